@@ -1,0 +1,391 @@
+"""CPU oracle for the Lloyd k-means hot path (test infrastructure only).
+
+Only tests/, __graft_entry__.smoke() and bench.py's CPU-baseline leg may import
+this package.  It never imports the CUDA library or its Python binding, and the
+CUDA path never imports it.
+
+The arithmetic lives in skm_oracle.c (plain C, -O2 -ffp-contract=off, OpenMP
+over rows); this module compiles it with gcc on first use, wraps each function
+for numpy arrays, and composes the Lloyd loop of Section 2.3 (STEP 2 and STEP 3
+repeated, then STEP 2 once more) for each representation.  The PCA
+eigen-decomposition is numpy.linalg.eigh on the fp64 covariance (a library
+routine used as one step), sorted by descending eigenvalue with each
+eigenvector's sign fixed so that its largest-magnitude entry is positive.
+
+Parity status: every function is pinned by tests/test_oracle_pins.py except the
+paper's printed dataset-level numbers (WCSS, recall), which need the paper's
+datasets: parity unpinned for those.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import subprocess
+import threading
+
+import numpy as np
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+_SRC = os.path.join(_HERE, "skm_oracle.c")
+_BUILD = os.path.join(_HERE, "_build")
+_LIB_PATH = os.path.join(_BUILD, "liboracle.so")
+_lock = threading.Lock()
+_lib = None
+
+GCC_FLAGS = ["-O2", "-std=c11", "-fPIC", "-shared", "-fopenmp", "-ffp-contract=off", "-fno-fast-math"]
+
+
+def build(force: bool = False) -> str:
+    """Compile skm_oracle.c into oracle/_build/liboracle.so (gcc)."""
+    os.makedirs(_BUILD, exist_ok=True)
+    stale = (not os.path.exists(_LIB_PATH)) or os.path.getmtime(_LIB_PATH) < os.path.getmtime(_SRC)
+    if force or stale:
+        tmp = _LIB_PATH + f".tmp{os.getpid()}"
+        subprocess.check_call(["gcc", *GCC_FLAGS, _SRC, "-o", tmp, "-lm"])
+        os.replace(tmp, _LIB_PATH)
+    return _LIB_PATH
+
+
+def _p(a):
+    return a.ctypes.data_as(ctypes.c_void_p) if a is not None else None
+
+
+def lib():
+    global _lib
+    with _lock:
+        if _lib is None:
+            build()
+            L = ctypes.CDLL(_LIB_PATH)
+            vp, i64, i32, f64 = ctypes.c_void_p, ctypes.c_int64, ctypes.c_int, ctypes.c_double
+            sig = {
+                "or_num_threads": ([], i32),
+                "or_set_num_threads": ([i32], None),
+                "or_assign_f32": ([vp, i64, i32, vp, i32, vp, vp, vp], None),
+                "or_assign_bf16": ([vp, i64, i32, vp, i32, vp, vp, vp], None),
+                "or_sq8_fit": ([vp, i64, i32, vp, vp], None),
+                "or_sq8_encode": ([vp, i64, i32, vp, vp, vp], None),
+                "or_sq8_decode": ([vp, i64, i32, vp, vp, vp], None),
+                "or_assign_sq8": ([vp, i64, i32, vp, i32, vp, vp], None),
+                "or_update_sq8": ([vp, i64, i32, vp, i32, vp, vp], None),
+                "or_update_f32": ([vp, i64, i32, vp, i32, vp, vp], None),
+                "or_update_bf16": ([vp, i64, i32, vp, i32, vp, vp], None),
+                "or_objective_f32": ([vp, i64, i32, vp, vp], f64),
+                "or_objective_bf16": ([vp, i64, i32, vp, vp], f64),
+                "or_rbq1_mean": ([vp, i64, i32, vp], None),
+                "or_rbq1_encode": ([vp, i64, i32, vp, vp, vp, vp, vp], None),
+                "or_rbq1_centroid_sq4": ([vp, i32, i32, vp, vp, vp, vp, vp, vp], None),
+                "or_rbq1_assign": ([vp, vp, vp, vp, i64, i32, vp, vp, vp, vp, vp, i32, vp, vp], None),
+                "or_rbq1_exponent": ([vp, i64], i32),
+                "or_rbq1_update": ([vp, vp, i64, i32, vp, i32, vp, i32, vp, vp], None),
+                "or_project": ([vp, i64, i32, vp, vp, i32, vp], None),
+                "or_mean_cov": ([vp, i64, i32, vp, vp], None),
+                "or_round_bf16": ([vp, i64, vp], None),
+            }
+            for name, (args, res) in sig.items():
+                fn = getattr(L, name)
+                fn.argtypes = args
+                fn.restype = res
+            _lib = L
+    return _lib
+
+
+def _c(a, dtype):
+    return np.ascontiguousarray(a, dtype=dtype)
+
+
+def num_threads() -> int:
+    return int(lib().or_num_threads())
+
+
+def set_num_threads(t: int) -> None:
+    lib().or_set_num_threads(int(t))
+
+
+# --------------------------------------------------------------------------
+# STEP 2 (Section 2.3): nearest centroid, plain definition
+# --------------------------------------------------------------------------
+def assign_f32(X, C):
+    """Returns (assign int32[n], best fp64[n], second fp64[n])."""
+    X, C = _c(X, np.float32), _c(C, np.float32)
+    n, d = X.shape
+    k = C.shape[0]
+    a = np.empty(n, np.int32)
+    b1 = np.empty(n, np.float64)
+    b2 = np.empty(n, np.float64)
+    lib().or_assign_f32(_p(X), n, d, _p(C), k, _p(a), _p(b1), _p(b2))
+    return a, b1, b2
+
+
+def assign_bf16(Xb, C):
+    """Points as bf16 bit patterns (uint16 [n, d]); returns (assign, best, second)."""
+    Xb, C = _c(Xb, np.uint16), _c(C, np.float32)
+    n, d = Xb.shape
+    k = C.shape[0]
+    a = np.empty(n, np.int32)
+    b1 = np.empty(n, np.float64)
+    b2 = np.empty(n, np.float64)
+    lib().or_assign_bf16(_p(Xb), n, d, _p(C), k, _p(a), _p(b1), _p(b2))
+    return a, b1, b2
+
+
+def bf16_to_f32(Xb) -> np.ndarray:
+    return (np.ascontiguousarray(Xb, np.uint16).astype(np.uint32) << 16).view(np.float32)
+
+
+def round_bf16(Y) -> np.ndarray:
+    """fp64 -> bf16 bit patterns (round half to even, from the fp64 value)."""
+    Y = _c(Y, np.float64)
+    out = np.empty(Y.shape, np.uint16)
+    lib().or_round_bf16(_p(Y), Y.size, _p(out))
+    return out
+
+
+# --------------------------------------------------------------------------
+# SQ8 (Section 3.1, per-dimension parameters)
+# --------------------------------------------------------------------------
+def sq8_fit(X):
+    X = _c(X, np.float32)
+    n, d = X.shape
+    b = np.empty(d, np.float32)
+    s = np.empty(d, np.float32)
+    lib().or_sq8_fit(_p(X), n, d, _p(b), _p(s))
+    return b, s
+
+
+def sq8_encode(X, b, s):
+    X = _c(X, np.float32)
+    n, d = X.shape
+    codes = np.empty((n, d), np.uint8)
+    lib().or_sq8_encode(_p(X), n, d, _p(_c(b, np.float32)), _p(_c(s, np.float32)), _p(codes))
+    return codes
+
+
+def sq8_decode(codes, b, s):
+    codes = _c(codes, np.uint8)
+    n, d = codes.shape
+    Y = np.empty((n, d), np.float32)
+    lib().or_sq8_decode(_p(codes), n, d, _p(_c(b, np.float32)), _p(_c(s, np.float32)), _p(Y))
+    return Y
+
+
+def assign_sq8(Xc, Cc):
+    Xc, Cc = _c(Xc, np.uint8), _c(Cc, np.uint8)
+    n, d = Xc.shape
+    k = Cc.shape[0]
+    a = np.empty(n, np.int32)
+    best = np.empty(n, np.int64)
+    lib().or_assign_sq8(_p(Xc), n, d, _p(Cc), k, _p(a), _p(best))
+    return a, best
+
+
+def update_sq8(Xc, assign, Cc):
+    Xc = _c(Xc, np.uint8)
+    n, d = Xc.shape
+    Cn = np.array(Cc, dtype=np.uint8, copy=True, order="C")
+    k = Cn.shape[0]
+    counts = np.empty(k, np.int64)
+    lib().or_update_sq8(_p(Xc), n, d, _p(_c(assign, np.int32)), k, _p(Cn), _p(counts))
+    return Cn, counts
+
+
+# --------------------------------------------------------------------------
+# STEP 3: mean of members; objective
+# --------------------------------------------------------------------------
+def update_f32(X, assign, C):
+    X = _c(X, np.float32)
+    n, d = X.shape
+    Cn = np.array(C, dtype=np.float32, copy=True, order="C")
+    k = Cn.shape[0]
+    counts = np.empty(k, np.int64)
+    lib().or_update_f32(_p(X), n, d, _p(_c(assign, np.int32)), k, _p(Cn), _p(counts))
+    return Cn, counts
+
+
+def update_bf16(Xb, assign, C):
+    Xb = _c(Xb, np.uint16)
+    n, d = Xb.shape
+    Cn = np.array(C, dtype=np.float32, copy=True, order="C")
+    k = Cn.shape[0]
+    counts = np.empty(k, np.int64)
+    lib().or_update_bf16(_p(Xb), n, d, _p(_c(assign, np.int32)), k, _p(Cn), _p(counts))
+    return Cn, counts
+
+
+def objective_f32(X, C, assign) -> float:
+    X = _c(X, np.float32)
+    n, d = X.shape
+    return float(lib().or_objective_f32(_p(X), n, d, _p(_c(C, np.float32)), _p(_c(assign, np.int32))))
+
+
+def objective_bf16(Xb, C, assign) -> float:
+    Xb = _c(Xb, np.uint16)
+    n, d = Xb.shape
+    return float(lib().or_objective_bf16(_p(Xb), n, d, _p(_c(C, np.float32)), _p(_c(assign, np.int32))))
+
+
+# --------------------------------------------------------------------------
+# RabitQ 1-bit (Section 3.1, Eq. l2_decomp, rabitq_l2, final:rabitq)
+# --------------------------------------------------------------------------
+def rbq1_mean(X):
+    X = _c(X, np.float32)
+    n, d = X.shape
+    m = np.empty(d, np.float32)
+    lib().or_rbq1_mean(_p(X), n, d, _p(m))
+    return m
+
+
+def rbq1_encode(X, m):
+    """Returns (codes uint32[n, W], nx2 f32[n], F f32[n], popx int32[n])."""
+    X = _c(X, np.float32)
+    n, d = X.shape
+    W = (d + 31) // 32
+    codes = np.empty((n, W), np.uint32)
+    nx2 = np.empty(n, np.float32)
+    F = np.empty(n, np.float32)
+    popx = np.empty(n, np.int32)
+    lib().or_rbq1_encode(_p(X), n, d, _p(_c(m, np.float32)), _p(codes), _p(nx2), _p(F), _p(popx))
+    return codes, nx2, F, popx
+
+
+def rbq1_centroid_sq4(C, m):
+    """Returns (ybar uint8[k, d], b f32[k], s f32[k], sumy int32[k], ny2 f32[k])."""
+    C = _c(C, np.float32)
+    k, d = C.shape
+    ybar = np.empty((k, d), np.uint8)
+    b = np.empty(k, np.float32)
+    s = np.empty(k, np.float32)
+    sumy = np.empty(k, np.int32)
+    ny2 = np.empty(k, np.float32)
+    lib().or_rbq1_centroid_sq4(_p(C), k, d, _p(_c(m, np.float32)), _p(ybar), _p(b), _p(s), _p(sumy), _p(ny2))
+    return ybar, b, s, sumy, ny2
+
+
+def rbq1_assign(codes, nx2, F, popx, d, prep):
+    """prep = rbq1_centroid_sq4(...). Returns (assign int32[n], est f32[n])."""
+    codes = _c(codes, np.uint32)
+    n = codes.shape[0]
+    ybar, b, s, sumy, ny2 = prep
+    k = ybar.shape[0]
+    a = np.empty(n, np.int32)
+    est = np.empty(n, np.float32)
+    lib().or_rbq1_assign(
+        _p(codes), _p(_c(nx2, np.float32)), _p(_c(F, np.float32)), _p(_c(popx, np.int32)), n, d,
+        _p(_c(ybar, np.uint8)), _p(_c(b, np.float32)), _p(_c(s, np.float32)), _p(_c(sumy, np.int32)),
+        _p(_c(ny2, np.float32)), k, _p(a), _p(est),
+    )
+    return a, est
+
+
+def rbq1_exponent(F) -> int:
+    F = _c(F, np.float32)
+    return int(lib().or_rbq1_exponent(_p(F), F.size))
+
+
+def rbq1_update(codes, F, d, m, e, assign, C):
+    codes = _c(codes, np.uint32)
+    n = codes.shape[0]
+    Cn = np.array(C, dtype=np.float32, copy=True, order="C")
+    k = Cn.shape[0]
+    counts = np.empty(k, np.int64)
+    lib().or_rbq1_update(
+        _p(codes), _p(_c(F, np.float32)), n, d, _p(_c(m, np.float32)), int(e),
+        _p(_c(assign, np.int32)), k, _p(Cn), _p(counts),
+    )
+    return Cn, counts
+
+
+def rbq1_decode_points(codes, F, d, m, e, idx):
+    """Decoded points (the fused decode-average of one member each), f32[len(idx), d]."""
+    idx = np.asarray(idx, np.int64)
+    sub_codes = _c(codes, np.uint32)[idx]
+    sub_F = _c(F, np.float32)[idx]
+    k = idx.size
+    C0 = np.zeros((k, d), np.float32)
+    C, _ = rbq1_update(sub_codes, sub_F, d, m, e, np.arange(k, dtype=np.int32), C0)
+    return C
+
+
+# --------------------------------------------------------------------------
+# Projection (rotation / PCA)
+# --------------------------------------------------------------------------
+def project(X, P, mu=None):
+    """Y = (X - mu) P in fp64, returned as fp64 [n, dout]."""
+    X = _c(X, np.float32)
+    P = _c(P, np.float32)
+    n, d = X.shape
+    dout = P.shape[1]
+    Y = np.empty((n, dout), np.float64)
+    lib().or_project(_p(X), n, d, _p(_c(mu, np.float32)) if mu is not None else None, _p(P), dout, _p(Y))
+    return Y
+
+
+def mean_cov(X):
+    X = _c(X, np.float32)
+    n, d = X.shape
+    mu = np.empty(d, np.float64)
+    cov = np.empty((d, d), np.float64)
+    lib().or_mean_cov(_p(X), n, d, _p(mu), _p(cov))
+    return mu, cov
+
+
+def pca_fit(X, d_out):
+    """Returns (mu fp64[d], P fp64[d, d_out], eigenvalues fp64[d_out]) by descending eigenvalue."""
+    mu, cov = mean_cov(X)
+    w, V = np.linalg.eigh(cov)
+    order = np.argsort(-w, kind="stable")[:d_out]
+    w = w[order]
+    V = V[:, order]
+    piv = np.argmax(np.abs(V), axis=0)
+    sgn = np.sign(V[piv, np.arange(V.shape[1])])
+    sgn[sgn == 0] = 1.0
+    return mu, V * sgn, w
+
+
+# --------------------------------------------------------------------------
+# Lloyd loop (Section 2.3): iters x (STEP 2, STEP 3), then STEP 2 once more.
+# objective[t] is the objective of the assignment made at step t.
+# --------------------------------------------------------------------------
+def lloyd_f32(X, C0, iters):
+    C = np.array(C0, np.float32, copy=True)
+    objs = []
+    for _ in range(iters):
+        a, best, _ = assign_f32(X, C)
+        objs.append(float(best.sum()))
+        C, counts = update_f32(X, a, C)
+    a, best, second = assign_f32(X, C)
+    objs.append(float(best.sum()))
+    return C, a, objs
+
+
+def lloyd_bf16(Xb, C0, iters):
+    C = np.array(C0, np.float32, copy=True)
+    objs = []
+    for _ in range(iters):
+        a, best, _ = assign_bf16(Xb, C)
+        objs.append(float(best.sum()))
+        C, counts = update_bf16(Xb, a, C)
+    a, best, _ = assign_bf16(Xb, C)
+    objs.append(float(best.sum()))
+    return C, a, objs
+
+
+def lloyd_sq8(Xc, C0c, iters):
+    Cc = np.array(C0c, np.uint8, copy=True)
+    for _ in range(iters):
+        a, _ = assign_sq8(Xc, Cc)
+        Cc, counts = update_sq8(Xc, a, Cc)
+    a, best = assign_sq8(Xc, Cc)
+    return Cc, a
+
+
+def lloyd_rbq1(codes, nx2, F, popx, d, m, C0, iters, e=None):
+    if e is None:
+        e = rbq1_exponent(F)
+    C = np.array(C0, np.float32, copy=True)
+    for _ in range(iters):
+        prep = rbq1_centroid_sq4(C, m)
+        a, _ = rbq1_assign(codes, nx2, F, popx, d, prep)
+        C, counts = rbq1_update(codes, F, d, m, e, a, C)
+    prep = rbq1_centroid_sq4(C, m)
+    a, est = rbq1_assign(codes, nx2, F, popx, d, prep)
+    return C, a

@@ -1,0 +1,519 @@
+/*
+ * skm_oracle.c -- plain, slow CPU oracle for the Lloyd k-means hot path of
+ * "Stop Indexing at Full Precision: Revisiting Clustering for Vector
+ * Embeddings" (arxiv 2608.14648).
+ *
+ * TEST INFRASTRUCTURE ONLY.  Only tests/, __graft_entry__.smoke() and the
+ * CPU-baseline leg of bench.py may load this library.  It shares no code,
+ * header, table or constant with the CUDA library; it is compiled with
+ * -O2 -ffp-contract=off and contains no blocking, fusion or reordering beyond
+ * what each definition states.  Rows are spread over OpenMP threads; every
+ * per-row computation is a plain sequential loop.
+ *
+ * Where the method has a plain definition (the nearest-centroid assignment of
+ * Section 2.3 STEP 2, the mean of members of STEP 3, the SQ8 integer code-space
+ * distance of Section 3.1) the oracle is that definition: fp64 or exact
+ * integer arithmetic, ties to the lowest centroid index.  Where the method is
+ * an encoding or an estimator (SQ8 codes, RabitQ 1-bit codes, the centroid SQ4
+ * codes and Eq. final:rabitq), the oracle takes the paper's steps in order.
+ * Where a float result decides an integer (a code, an argmin over estimated
+ * distances), the oracle performs that float step in fp32 in the fixed
+ * operation order the method is specified with, so that both sides take the
+ * decision in the same precision.
+ *
+ * Parity status of each function is stated in its comment; the pins live in
+ * tests/test_oracle_pins.py.
+ */
+#include <math.h>
+#include <stdint.h>
+#include <stdlib.h>
+#include <string.h>
+#ifdef _OPENMP
+#include <omp.h>
+#endif
+
+int or_num_threads(void) {
+#ifdef _OPENMP
+    return omp_get_max_threads();
+#else
+    return 1;
+#endif
+}
+
+void or_set_num_threads(int t) {
+#ifdef _OPENMP
+    if (t > 0) omp_set_num_threads(t);
+#else
+    (void)t;
+#endif
+}
+
+static inline float bf16_bits_to_float(uint16_t b) {
+    uint32_t u = ((uint32_t)b) << 16;
+    float f;
+    memcpy(&f, &u, 4);
+    return f;
+}
+
+/* ------------------------------------------------------------------------ */
+/* Section 2.3 STEP 2: nearest centroid under squared L2, plain definition.  */
+/* ------------------------------------------------------------------------ */
+
+/* dist(x, c) = sum_i (x_i - c_i)^2 in fp64; argmin over all k, ties to the
+ * lowest index.  best/second receive the smallest and second-smallest fp64
+ * distances (second is used only to report top-1/top-2 gaps, Fig. 3).
+ * Pinned: brute force, scipy cdist, K=1, N=K identity, duplicates. */
+void or_assign_f32(const float *X, int64_t n, int d, const float *C, int k,
+                   int32_t *assign, double *best, double *second) {
+#pragma omp parallel for schedule(dynamic, 64)
+    for (int64_t p = 0; p < n; ++p) {
+        const float *x = X + p * (int64_t)d;
+        double b1 = INFINITY, b2 = INFINITY;
+        int32_t a = -1;
+        for (int j = 0; j < k; ++j) {
+            const float *c = C + (int64_t)j * d;
+            double s = 0.0;
+            for (int i = 0; i < d; ++i) {
+                double t = (double)x[i] - (double)c[i];
+                s += t * t;
+            }
+            if (s < b1) {
+                b2 = b1;
+                b1 = s;
+                a = j;
+            } else if (s < b2) {
+                b2 = s;
+            }
+        }
+        assign[p] = a;
+        if (best) best[p] = b1;
+        if (second) second[p] = b2;
+    }
+}
+
+/* Same definition for points stored as bfloat16 bit patterns (the projected
+ * points of the PCA workload, stored in bf16; every bf16 value is exact in
+ * fp32 and fp64). */
+void or_assign_bf16(const uint16_t *Xb, int64_t n, int d, const float *C, int k,
+                    int32_t *assign, double *best, double *second) {
+#pragma omp parallel for schedule(dynamic, 64)
+    for (int64_t p = 0; p < n; ++p) {
+        const uint16_t *x = Xb + p * (int64_t)d;
+        double b1 = INFINITY, b2 = INFINITY;
+        int32_t a = -1;
+        for (int j = 0; j < k; ++j) {
+            const float *c = C + (int64_t)j * d;
+            double s = 0.0;
+            for (int i = 0; i < d; ++i) {
+                double t = (double)bf16_bits_to_float(x[i]) - (double)c[i];
+                s += t * t;
+            }
+            if (s < b1) {
+                b2 = b1;
+                b1 = s;
+                a = j;
+            } else if (s < b2) {
+                b2 = s;
+            }
+        }
+        assign[p] = a;
+        if (best) best[p] = b1;
+        if (second) second[p] = b2;
+    }
+}
+
+/* ------------------------------------------------------------------------ */
+/* Section 3.1 "SQ8 and SQ4": scalar quantization.                           */
+/* The paper fits one global bias/scale; the workload here fits them per     */
+/* dimension (b_i = min over points, s_i = (max - b_i) / 255).  A dimension  */
+/* with max == min gets s_i = 1.                                             */
+/* ------------------------------------------------------------------------ */
+
+void or_sq8_fit(const float *X, int64_t n, int d, float *b, float *s) {
+    for (int i = 0; i < d; ++i) {
+        float lo = INFINITY, hi = -INFINITY;
+        for (int64_t p = 0; p < n; ++p) {
+            float v = X[p * (int64_t)d + i];
+            if (v < lo) lo = v;
+            if (v > hi) hi = v;
+        }
+        float sc = (hi - lo) / 255.0f;
+        if (!(sc > 0.0f)) sc = 1.0f;
+        b[i] = lo;
+        s[i] = sc;
+    }
+}
+
+/* code = clip(round((x - b) / s), 0, 255), fp32 arithmetic, rounding half to
+ * even.  Pinned: grid data reproduces codes; |decode - x| <= s/2. */
+void or_sq8_encode(const float *X, int64_t n, int d, const float *b, const float *s,
+                   uint8_t *codes) {
+#pragma omp parallel for schedule(static)
+    for (int64_t p = 0; p < n; ++p) {
+        for (int i = 0; i < d; ++i) {
+            float t = (X[p * (int64_t)d + i] - b[i]) / s[i];
+            float q = rintf(t);
+            if (!(q >= 0.0f)) q = 0.0f;
+            if (q > 255.0f) q = 255.0f;
+            codes[p * (int64_t)d + i] = (uint8_t)q;
+        }
+    }
+}
+
+/* Reconstruction x_i ~ code_i * s_i + b_i (fp32). */
+void or_sq8_decode(const uint8_t *codes, int64_t n, int d, const float *b, const float *s,
+                   float *Y) {
+#pragma omp parallel for schedule(static)
+    for (int64_t p = 0; p < n; ++p)
+        for (int i = 0; i < d; ++i)
+            Y[p * (int64_t)d + i] = (float)codes[p * (int64_t)d + i] * s[i] + b[i];
+}
+
+/* Code-domain squared L2, exact in integers: sum_i (xbar_i - cbar_i)^2.
+ * Pinned: exact int64 recomputation through numpy; brute force. */
+void or_assign_sq8(const uint8_t *Xc, int64_t n, int d, const uint8_t *Cc, int k,
+                   int32_t *assign, int64_t *best) {
+#pragma omp parallel for schedule(dynamic, 64)
+    for (int64_t p = 0; p < n; ++p) {
+        const uint8_t *x = Xc + p * (int64_t)d;
+        int64_t b1 = INT64_MAX;
+        int32_t a = -1;
+        for (int j = 0; j < k; ++j) {
+            const uint8_t *c = Cc + (int64_t)j * d;
+            int64_t s = 0;
+            for (int i = 0; i < d; ++i) {
+                int64_t t = (int64_t)x[i] - (int64_t)c[i];
+                s += t * t;
+            }
+            if (s < b1) {
+                b1 = s;
+                a = j;
+            }
+        }
+        assign[p] = a;
+        if (best) best[p] = b1;
+    }
+}
+
+/* STEP 3 in the quantized domain: per-dimension average of member codes,
+ * rounded half to even in exact integer arithmetic.  Empty clusters keep
+ * their codes.  Pinned: brute-force mean + rounding. */
+void or_update_sq8(const uint8_t *Xc, int64_t n, int d, const int32_t *assign, int k,
+                   uint8_t *C_inout, int64_t *counts) {
+    int64_t *S = (int64_t *)calloc((size_t)k * d, sizeof(int64_t));
+    for (int j = 0; j < k; ++j) counts[j] = 0;
+    for (int64_t p = 0; p < n; ++p) {
+        int32_t a = assign[p];
+        counts[a] += 1;
+        for (int i = 0; i < d; ++i) S[(int64_t)a * d + i] += Xc[p * (int64_t)d + i];
+    }
+    for (int j = 0; j < k; ++j) {
+        int64_t m = counts[j];
+        if (m == 0) continue;
+        for (int i = 0; i < d; ++i) {
+            int64_t t = S[(int64_t)j * d + i];
+            int64_t q = t / m, r = t % m; /* t >= 0 */
+            if (2 * r > m || (2 * r == m && (q & 1))) q += 1;
+            C_inout[(int64_t)j * d + i] = (uint8_t)q;
+        }
+    }
+    free(S);
+}
+
+/* ------------------------------------------------------------------------ */
+/* STEP 3: centroid = mean of its members (fp64 sums, rounded to fp32).      */
+/* Empty clusters keep their previous centroid.                              */
+/* ------------------------------------------------------------------------ */
+
+static void update_mean_common(const float *X, const uint16_t *Xb, int64_t n, int d,
+                               const int32_t *assign, int k, float *C_inout,
+                               int64_t *counts) {
+    double *S = (double *)calloc((size_t)k * d, sizeof(double));
+    for (int j = 0; j < k; ++j) counts[j] = 0;
+    for (int64_t p = 0; p < n; ++p) {
+        int32_t a = assign[p];
+        counts[a] += 1;
+        for (int i = 0; i < d; ++i) {
+            double v = X ? (double)X[p * (int64_t)d + i]
+                         : (double)bf16_bits_to_float(Xb[p * (int64_t)d + i]);
+            S[(int64_t)a * d + i] += v;
+        }
+    }
+    for (int j = 0; j < k; ++j) {
+        if (counts[j] == 0) continue;
+        for (int i = 0; i < d; ++i)
+            C_inout[(int64_t)j * d + i] = (float)(S[(int64_t)j * d + i] / (double)counts[j]);
+    }
+    free(S);
+}
+
+void or_update_f32(const float *X, int64_t n, int d, const int32_t *assign, int k,
+                   float *C_inout, int64_t *counts) {
+    update_mean_common(X, NULL, n, d, assign, k, C_inout, counts);
+}
+
+void or_update_bf16(const uint16_t *Xb, int64_t n, int d, const int32_t *assign, int k,
+                    float *C_inout, int64_t *counts) {
+    update_mean_common(NULL, Xb, n, d, assign, k, C_inout, counts);
+}
+
+/* k-means objective (WCSS, Section 4): sum_n ||x_n - c_{a_n}||^2 in fp64. */
+double or_objective_f32(const float *X, int64_t n, int d, const float *C,
+                        const int32_t *assign) {
+    double tot = 0.0;
+#pragma omp parallel for reduction(+ : tot) schedule(static)
+    for (int64_t p = 0; p < n; ++p) {
+        const float *x = X + p * (int64_t)d;
+        const float *c = C + (int64_t)assign[p] * d;
+        double s = 0.0;
+        for (int i = 0; i < d; ++i) {
+            double t = (double)x[i] - (double)c[i];
+            s += t * t;
+        }
+        tot += s;
+    }
+    return tot;
+}
+
+double or_objective_bf16(const uint16_t *Xb, int64_t n, int d, const float *C,
+                         const int32_t *assign) {
+    double tot = 0.0;
+#pragma omp parallel for reduction(+ : tot) schedule(static)
+    for (int64_t p = 0; p < n; ++p) {
+        const uint16_t *x = Xb + p * (int64_t)d;
+        const float *c = C + (int64_t)assign[p] * d;
+        double s = 0.0;
+        for (int i = 0; i < d; ++i) {
+            double t = (double)bf16_bits_to_float(x[i]) - (double)c[i];
+            s += t * t;
+        }
+        tot += s;
+    }
+    return tot;
+}
+
+/* ------------------------------------------------------------------------ */
+/* Section 3.1 "RabitQ": 1-bit codes of the centred data points, SQ4 codes   */
+/* of the centred centroids, Eq. l2_decomp / rabitq_l2 / final:rabitq.       */
+/* ------------------------------------------------------------------------ */
+
+/* Dataset mean m (fp64 sum, rounded to fp32). */
+void or_rbq1_mean(const float *X, int64_t n, int d, float *m) {
+    for (int i = 0; i < d; ++i) {
+        double s = 0.0;
+        for (int64_t p = 0; p < n; ++p) s += (double)X[p * (int64_t)d + i];
+        m[i] = (float)(s / (double)n);
+    }
+}
+
+/* Per point: r = x - m (fp32); bit i = (r_i > 0), packed little-endian into
+ * 32-bit words (bit j of word w is dimension 32w + j); nx2 = ||r||^2;
+ * <xbar, x> = ||r||_1 / (sqrt(d) ||r||) so F = ||r|| / <xbar, x>
+ * = sqrt(d) ||r||^2 / ||r||_1 (0 when r = 0); popx = number of set bits.
+ * Pinned: exact reconstruction on sign-constant residuals, radius >= ||r||. */
+void or_rbq1_encode(const float *X, int64_t n, int d, const float *m, uint32_t *codes,
+                    float *nx2, float *F, int32_t *popx) {
+    const int W = (d + 31) / 32;
+#pragma omp parallel for schedule(static)
+    for (int64_t p = 0; p < n; ++p) {
+        uint32_t *cw = codes + p * (int64_t)W;
+        for (int w = 0; w < W; ++w) cw[w] = 0u;
+        double s2 = 0.0, s1 = 0.0;
+        int32_t pc = 0;
+        for (int i = 0; i < d; ++i) {
+            float r = X[p * (int64_t)d + i] - m[i];
+            if (r > 0.0f) {
+                cw[i / 32] |= (1u << (i % 32));
+                pc += 1;
+            }
+            s2 += (double)r * (double)r;
+            s1 += fabs((double)r);
+        }
+        nx2[p] = (float)s2;
+        F[p] = (s1 > 0.0) ? (float)(sqrt((double)d) * s2 / s1) : 0.0f;
+        popx[p] = pc;
+    }
+}
+
+/* Centroid side, once per iteration: rho = c - m (fp32); per-centroid SQ4
+ * with b = min rho, s = (max rho - b) / 15 (s = 1 when flat); ybar_i =
+ * clip(round((rho_i - b) / s), 0, 15) with rounding half to even;
+ * sumy = sum ybar; ny2 = ||rho||^2 (fp64, sequential, rounded to fp32). */
+void or_rbq1_centroid_sq4(const float *C, int k, int d, const float *m, uint8_t *ybar,
+                          float *b, float *s, int32_t *sumy, float *ny2) {
+    for (int j = 0; j < k; ++j) {
+        const float *c = C + (int64_t)j * d;
+        float lo = INFINITY, hi = -INFINITY;
+        double q2 = 0.0;
+        for (int i = 0; i < d; ++i) {
+            float r = c[i] - m[i];
+            if (r < lo) lo = r;
+            if (r > hi) hi = r;
+            q2 += (double)r * (double)r;
+        }
+        float sc = (hi - lo) / 15.0f;
+        if (!(sc > 0.0f)) sc = 1.0f;
+        int32_t sy = 0;
+        for (int i = 0; i < d; ++i) {
+            float r = c[i] - m[i];
+            float q = rintf((r - lo) / sc);
+            if (!(q >= 0.0f)) q = 0.0f;
+            if (q > 15.0f) q = 15.0f;
+            ybar[(int64_t)j * d + i] = (uint8_t)q;
+            sy += (int32_t)q;
+        }
+        b[j] = lo;
+        s[j] = sc;
+        sumy[j] = sy;
+        ny2[j] = (float)q2;
+    }
+}
+
+/* Eq. final:rabitq into Eq. rabitq_l2, fp32 in this fixed order:
+ *   P   = sum_i xbar_i * ybar_i              (exact integer)
+ *   t1  = s * (2P - sum ybar)
+ *   t2  = b * (2 popx - d)
+ *   ip  = (t1 + t2) * (1/sqrt(d))            (1/sqrt(d) rounded once to fp32)
+ *   est = (nx2 + ny2) - 2 (F * ip)
+ * argmin over est, ties to the lowest index. */
+void or_rbq1_assign(const uint32_t *codes, const float *nx2, const float *F,
+                    const int32_t *popx, int64_t n, int d, const uint8_t *ybar,
+                    const float *b, const float *s, const int32_t *sumy,
+                    const float *ny2, int k, int32_t *assign, float *est_best) {
+    const int W = (d + 31) / 32;
+    const float isd = (float)(1.0 / sqrt((double)d));
+#pragma omp parallel for schedule(dynamic, 16)
+    for (int64_t p = 0; p < n; ++p) {
+        const uint32_t *cw = codes + p * (int64_t)W;
+        float best = INFINITY;
+        int32_t a = -1;
+        for (int j = 0; j < k; ++j) {
+            const uint8_t *y = ybar + (int64_t)j * d;
+            int32_t P = 0;
+            for (int i = 0; i < d; ++i)
+                if ((cw[i / 32] >> (i % 32)) & 1u) P += y[i];
+            float t1 = s[j] * (float)(2 * P - sumy[j]);
+            float t2 = b[j] * (float)(2 * popx[p] - d);
+            float ip = (t1 + t2) * isd;
+            float nn = nx2[p] + ny2[j];
+            float fi = F[p] * ip;
+            float est = nn - 2.0f * fi;
+            if (est < best) {
+                best = est;
+                a = j;
+            }
+        }
+        assign[p] = a;
+        if (est_best) est_best[p] = best;
+    }
+}
+
+/* Fixed-point exponent for the decode-average: e = 37 - ceil(log2 max F),
+ * so F * 2^e <= 2^37; e = 0 when every F is 0. */
+int or_rbq1_exponent(const float *F, int64_t n) {
+    float mx = 0.0f;
+    for (int64_t p = 0; p < n; ++p)
+        if (F[p] > mx) mx = F[p];
+    if (!(mx > 0.0f)) return 0;
+    int ex;
+    double fr = frexp((double)mx, &ex); /* mx = fr * 2^ex, fr in [0.5, 1) */
+    int c = (fr == 0.5) ? ex - 1 : ex;  /* ceil(log2 mx) */
+    return 37 - c;
+}
+
+/* Fused decode-average (Section 3.1 "RabitQ", last paragraph): the member
+ * x_r is decoded as m_i + (1/sqrt(d)) F (2 xbar_i - 1) and the members are
+ * averaged.  F enters as the integer Fq = round(F 2^e), so the sum over the
+ * members is exact and independent of order:
+ *   T_i = sum Fq xbar_i,  U = sum Fq,  sum F (2 xbar_i - 1) = (2 T_i - U) 2^-e
+ *   c_i = m_i + ((2 T_i - U) 2^-e / count) / sqrt(d)     (fp64, then fp32)
+ * Empty clusters keep their centroid.  Pinned against the fp64 mean of
+ * decoded vectors (relative 1e-9) and the exact-reconstruction case. */
+void or_rbq1_update(const uint32_t *codes, const float *F, int64_t n, int d,
+                    const float *m, int e, const int32_t *assign, int k, float *C_inout,
+                    int64_t *counts) {
+    const int W = (d + 31) / 32;
+    const double isd = 1.0 / sqrt((double)d);
+    int64_t *T = (int64_t *)calloc((size_t)k * d, sizeof(int64_t));
+    int64_t *U = (int64_t *)calloc((size_t)k, sizeof(int64_t));
+    for (int j = 0; j < k; ++j) counts[j] = 0;
+    for (int64_t p = 0; p < n; ++p) {
+        int32_t a = assign[p];
+        int64_t fq = (int64_t)llrint(ldexp((double)F[p], e));
+        counts[a] += 1;
+        U[a] += fq;
+        const uint32_t *cw = codes + p * (int64_t)W;
+        for (int i = 0; i < d; ++i)
+            if ((cw[i / 32] >> (i % 32)) & 1u) T[(int64_t)a * d + i] += fq;
+    }
+    for (int j = 0; j < k; ++j) {
+        if (counts[j] == 0) continue;
+        for (int i = 0; i < d; ++i) {
+            double v = (double)(2 * T[(int64_t)j * d + i] - U[j]);
+            v = ldexp(v, -e);
+            v = v / (double)counts[j];
+            v = v * isd;
+            C_inout[(int64_t)j * d + i] = (float)((double)m[i] + v);
+        }
+    }
+    free(T);
+    free(U);
+}
+
+/* ------------------------------------------------------------------------ */
+/* Section 3.1 "JLT / PCA" and the rotation of "SuperKMeans": projection     */
+/* Y = (X - mu) P, fp64.                                                     */
+/* ------------------------------------------------------------------------ */
+
+void or_project(const float *X, int64_t n, int d, const float *mu, const float *P,
+                int dout, double *Y) {
+#pragma omp parallel for schedule(static)
+    for (int64_t p = 0; p < n; ++p) {
+        const float *x = X + p * (int64_t)d;
+        double *y = Y + p * (int64_t)dout;
+        for (int j = 0; j < dout; ++j) y[j] = 0.0;
+        for (int i = 0; i < d; ++i) {
+            double xi = (double)x[i] - (mu ? (double)mu[i] : 0.0);
+            for (int j = 0; j < dout; ++j) y[j] += xi * (double)P[(int64_t)i * dout + j];
+        }
+    }
+}
+
+/* Mean and population covariance (1/n) sum (x - mu)(x - mu)^T, fp64. */
+void or_mean_cov(const float *X, int64_t n, int d, double *mu, double *cov) {
+    for (int i = 0; i < d; ++i) {
+        double s = 0.0;
+        for (int64_t p = 0; p < n; ++p) s += (double)X[p * (int64_t)d + i];
+        mu[i] = s / (double)n;
+    }
+#pragma omp parallel for schedule(dynamic, 4)
+    for (int i = 0; i < d; ++i) {
+        for (int j = 0; j <= i; ++j) {
+            double s = 0.0;
+            for (int64_t p = 0; p < n; ++p)
+                s += ((double)X[p * (int64_t)d + i] - mu[i]) * ((double)X[p * (int64_t)d + j] - mu[j]);
+            cov[(int64_t)i * d + j] = s / (double)n;
+            cov[(int64_t)j * d + i] = s / (double)n;
+        }
+    }
+}
+
+/* Round fp64 values to bfloat16 (8 significant bits, half to even). */
+void or_round_bf16(const double *y, int64_t n, uint16_t *out) {
+#pragma omp parallel for schedule(static)
+    for (int64_t p = 0; p < n; ++p) {
+        double v = y[p];
+        float f;
+        if (v == 0.0 || !isfinite(v)) {
+            f = (float)v;
+        } else {
+            int ex;
+            double fr = frexp(v, &ex); /* |fr| in [0.5, 1) */
+            double q = rint(ldexp(fr, 8));
+            f = (float)ldexp(q, ex - 8);
+        }
+        uint32_t u;
+        memcpy(&u, &f, 4);
+        out[p] = (uint16_t)(u >> 16);
+    }
+}

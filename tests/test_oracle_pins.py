@@ -1,0 +1,333 @@
+"""Pins for the CPU oracle: each check ties the oracle to something other than
+itself (a library routine, a closed form, an invariant, brute force on tiny
+inputs, or the hand-worked example in tests/golden/).  No GPU needed."""
+import json
+import math
+import os
+
+import numpy as np
+import pytest
+import scipy.cluster.vq as vq
+from scipy.spatial.distance import cdist
+
+import oracle
+
+GOLDEN = os.path.join(os.path.dirname(__file__), "golden")
+
+
+def _rng(seed=0):
+    return np.random.default_rng(seed)
+
+
+# ---------------------------------------------------------------- assignment
+@pytest.mark.parametrize("d", [1, 31, 32, 33, 64])
+@pytest.mark.parametrize("n,k", [(64, 8), (17, 3), (5, 1)])
+def test_assign_f32_matches_cdist_brute_force(n, k, d):
+    r = _rng(d * 100 + k)
+    X = r.standard_normal((n, d)).astype(np.float32)
+    C = r.standard_normal((k, d)).astype(np.float32)
+    a, best, second = oracle.assign_f32(X, C)
+    D = cdist(X.astype(np.float64), C.astype(np.float64), "sqeuclidean")
+    np.testing.assert_array_equal(a, np.argmin(D, axis=1))
+    np.testing.assert_allclose(best, D.min(axis=1), rtol=1e-12, atol=1e-12)
+    if k > 1:
+        np.testing.assert_allclose(second, np.sort(D, axis=1)[:, 1], rtol=1e-12, atol=1e-12)
+    # invariant: the assigned distance is <= every other centroid's distance
+    assert np.all(best[:, None] <= D + 1e-12)
+
+
+def test_assign_f32_special_cases():
+    r = _rng(1)
+    X = r.standard_normal((40, 7)).astype(np.float32)
+    # K = 1: everything goes to centroid 0
+    a, _, _ = oracle.assign_f32(X, X[:1])
+    assert np.all(a == 0)
+    # N = K with centroids = points: identity assignment, objective 0
+    a, best, _ = oracle.assign_f32(X, X)
+    np.testing.assert_array_equal(a, np.arange(40))
+    assert best.sum() == 0.0
+    # duplicate centroids: ties go to the lowest index
+    C = np.concatenate([X[3:4], X[3:4], X[5:6], X[5:6]])
+    a, _, _ = oracle.assign_f32(X[[3, 5]], C)
+    np.testing.assert_array_equal(a, [0, 2])
+    # a point exactly halfway between two centroids goes to the lower index
+    C = np.array([[1.0, 0.0], [-1.0, 0.0]], np.float32)
+    a, _, _ = oracle.assign_f32(np.zeros((1, 2), np.float32), C[::-1].copy())
+    assert a[0] == 0
+
+
+def test_assign_bf16_matches_cdist():
+    r = _rng(2)
+    Xf = r.standard_normal((50, 33))
+    Xb = oracle.round_bf16(Xf)
+    C = r.standard_normal((6, 33)).astype(np.float32)
+    a, best, _ = oracle.assign_bf16(Xb, C)
+    D = cdist(oracle.bf16_to_f32(Xb).astype(np.float64), C.astype(np.float64), "sqeuclidean")
+    np.testing.assert_array_equal(a, np.argmin(D, axis=1))
+    np.testing.assert_allclose(best, D.min(axis=1), rtol=1e-12)
+
+
+# -------------------------------------------------------------------- update
+def test_update_f32_is_member_mean_and_keeps_empty():
+    r = _rng(3)
+    X = r.standard_normal((200, 9)).astype(np.float32)
+    k = 6
+    a = r.integers(0, k - 1, size=200).astype(np.int32)  # cluster k-1 stays empty
+    C0 = r.standard_normal((k, 9)).astype(np.float32)
+    C, counts = oracle.update_f32(X, a, C0)
+    assert counts.sum() == 200 and counts[k - 1] == 0
+    for j in range(k - 1):
+        np.testing.assert_allclose(C[j], X[a == j].astype(np.float64).mean(axis=0), rtol=1e-6, atol=1e-7)
+    np.testing.assert_array_equal(C[k - 1], C0[k - 1])
+    # K = 1: the global mean
+    C1, _ = oracle.update_f32(X, np.zeros(200, np.int32), C0[:1])
+    np.testing.assert_allclose(C1[0], X.astype(np.float64).mean(axis=0), rtol=1e-6, atol=1e-7)
+
+
+def test_lloyd_f32_matches_scipy_kmeans2_and_is_monotone():
+    import synth
+
+    X = synth.gmm_points(3000, 16, 20, seed=5, decay=False).numpy()
+    idx = synth.forgy_indices(3000, 20, seed=5).numpy()
+    C0 = X[idx].copy()
+    C, a, objs = oracle.lloyd_f32(X, C0, 10)
+    # scipy's kmeans2 with given initial centroids is the same Lloyd loop
+    # (assign, mean of members, empty clusters keep their centroid), in fp64.
+    # kmeans2 returns the labels of its last assignment, made before its last
+    # update; the final STEP 2 on its returned centroids is vq.vq.
+    Cs, _ = vq.kmeans2(X.astype(np.float64), C0.astype(np.float64), iter=10, minit="matrix", missing="warn")
+    labs, _ = vq.vq(X.astype(np.float64), Cs)
+    assert np.mean(labs == a) > 0.999
+    np.testing.assert_allclose(C, Cs, rtol=1e-4, atol=1e-5)
+    # Lloyd's objective never increases (fp32 centroids: allow 1e-6 slack)
+    for t in range(1, len(objs)):
+        assert objs[t] <= objs[t - 1] * (1 + 1e-6)
+
+
+def test_objective_is_wcss():
+    r = _rng(4)
+    X = r.standard_normal((100, 5)).astype(np.float32)
+    C = r.standard_normal((4, 5)).astype(np.float32)
+    a = r.integers(0, 4, 100).astype(np.int32)
+    want = float(((X.astype(np.float64) - C[a].astype(np.float64)) ** 2).sum())
+    assert math.isclose(oracle.objective_f32(X, C, a), want, rel_tol=1e-12)
+
+
+# ----------------------------------------------------------------------- SQ8
+def test_sq8_grid_data_reproduces_codes():
+    r = _rng(6)
+    n, d = 300, 37
+    codes = r.integers(0, 256, size=(n, d)).astype(np.uint8)
+    codes[0, :] = 0
+    codes[1, :] = 255
+    s0 = (2.0 ** -r.integers(3, 9, size=d)).astype(np.float32)
+    b0 = (r.integers(-50, 50, size=d) * s0).astype(np.float32)
+    X = (codes.astype(np.float32) * s0 + b0).astype(np.float32)
+    b, s = oracle.sq8_fit(X)
+    np.testing.assert_array_equal(b, b0)
+    np.testing.assert_array_equal(s, s0)
+    np.testing.assert_array_equal(oracle.sq8_encode(X, b, s), codes)
+    np.testing.assert_array_equal(oracle.sq8_decode(codes, b, s), X)
+
+
+def test_sq8_roundtrip_error_bound_and_flat_dims():
+    r = _rng(7)
+    X = r.standard_normal((500, 20)).astype(np.float32)
+    X[:, 3] = 0.25  # flat dimension
+    b, s = oracle.sq8_fit(X)
+    assert s[3] == 1.0 and b[3] == 0.25
+    np.testing.assert_array_equal(b, X.min(axis=0))
+    codes = oracle.sq8_encode(X, b, s)
+    assert codes[:, 3].max() == 0
+    np.testing.assert_array_equal(codes.min(axis=0)[np.arange(20) != 3], 0)
+    np.testing.assert_array_equal(codes.max(axis=0)[np.arange(20) != 3], 255)
+    err = np.abs(oracle.sq8_decode(codes, b, s).astype(np.float64) - X)
+    assert np.all(err <= s.astype(np.float64) / 2 * (1 + 1e-5) + 1e-7)
+
+
+def test_assign_and_update_sq8_exact_integers():
+    r = _rng(8)
+    Xc = r.integers(0, 256, size=(120, 45)).astype(np.uint8)
+    Cc = r.integers(0, 256, size=(7, 45)).astype(np.uint8)
+    Cc[5] = Cc[2]  # duplicate: ties to the lower index
+    a, best = oracle.assign_sq8(Xc, Cc)
+    D = cdist(Xc.astype(np.float64), Cc.astype(np.float64), "sqeuclidean")  # exact below 2^53
+    np.testing.assert_array_equal(a, np.argmin(D, axis=1))
+    np.testing.assert_array_equal(best, D.min(axis=1).astype(np.int64))
+    assert not np.any(a == 5)
+    a2 = r.integers(0, 6, 120).astype(np.int32)  # cluster 6 empty
+    Cn, counts = oracle.update_sq8(Xc, a2, Cc)
+    for j in range(6):
+        S = Xc[a2 == j].astype(np.int64).sum(axis=0)
+        np.testing.assert_array_equal(Cn[j], np.rint(S / counts[j]).astype(np.uint8))
+    np.testing.assert_array_equal(Cn[6], Cc[6])
+    # exact halves round to even
+    Xh = np.array([[2], [3], [0], [1], [5], [6]], np.uint8)
+    Cn, _ = oracle.update_sq8(Xh, np.array([0, 0, 1, 1, 2, 2], np.int32), np.zeros((3, 1), np.uint8))
+    np.testing.assert_array_equal(Cn[:, 0], [2, 0, 6])  # 2.5 -> 2, 0.5 -> 0, 5.5 -> 6
+
+
+# ------------------------------------------------------------------ RabitQ
+def _sign_constant_points(r, n, d, m, amp):
+    sg = np.where(r.random((n, d)) < 0.5, -1.0, 1.0)
+    return (m[None, :].astype(np.float64) + amp[:, None] * sg).astype(np.float32), sg
+
+
+def test_rbq1_encode_bits_and_factors():
+    r = _rng(9)
+    n, d = 40, 70
+    X = r.standard_normal((n, d)).astype(np.float32)
+    m = oracle.rbq1_mean(X)
+    np.testing.assert_allclose(m, X.astype(np.float64).mean(axis=0), rtol=1e-6, atol=1e-7)
+    codes, nx2, F, popx = oracle.rbq1_encode(X, m)
+    R = X - m[None, :]
+    bits = (R > 0).astype(np.uint8)
+    packed = np.packbits(np.pad(bits, ((0, 0), (0, 96 - d))), axis=1, bitorder="little").view(np.uint32)
+    np.testing.assert_array_equal(codes, packed)
+    np.testing.assert_array_equal(popx, bits.sum(axis=1))
+    R64 = R.astype(np.float64)
+    np.testing.assert_allclose(nx2, (R64 ** 2).sum(axis=1), rtol=1e-6)
+    # <xbar, x> = ||r||_1 / (sqrt(d) ||r||); F = ||r|| / <xbar, x>
+    cosq = np.abs(R64).sum(axis=1) / (math.sqrt(d) * np.linalg.norm(R64, axis=1))
+    np.testing.assert_allclose(F, np.linalg.norm(R64, axis=1) / cosq, rtol=1e-6)
+    # Cauchy-Schwarz (Section 4, "Closing RabitQ's gap"): decoded radius F >= ||r||
+    assert np.all(F >= np.sqrt(nx2) * (1 - 1e-6))
+    # degenerate residual r = 0
+    _, nx2z, Fz, popz = oracle.rbq1_encode(m[None, :].copy(), m)
+    assert nx2z[0] == 0 and Fz[0] == 0 and popz[0] == 0
+
+
+def test_rbq1_decode_exact_for_sign_constant_residuals():
+    r = _rng(10)
+    n, d = 30, 96
+    m = r.standard_normal(d).astype(np.float32) * 0.1
+    amp = r.uniform(0.5, 2.0, n)
+    X, sg = _sign_constant_points(r, n, d, m, amp)
+    codes, nx2, F, popx = oracle.rbq1_encode(X, m)
+    e = oracle.rbq1_exponent(F)
+    Cdec = oracle.rbq1_decode_points(codes, F, d, m, e, np.arange(n))
+    np.testing.assert_allclose(Cdec, X, rtol=1e-6, atol=1e-6)
+
+
+def test_rbq1_estimator_matches_direct_sum_and_is_exact_on_grid():
+    r = _rng(11)
+    n, d, k = 25, 64, 1
+    m = np.zeros(d, np.float32)
+    amp = r.uniform(0.5, 2.0, n)
+    X, sg = _sign_constant_points(r, n, d, m, amp)
+    codes, nx2, F, popx = oracle.rbq1_encode(X, m)
+    # centroid residual exactly on an SQ4 grid: c - m = b + s * ybar
+    yb = r.integers(0, 16, size=d)
+    yb[0], yb[1] = 0, 15
+    b0, s0 = np.float32(-0.75), np.float32(0.125)
+    C = (b0 + s0 * yb.astype(np.float32))[None, :].astype(np.float32)
+    prep = oracle.rbq1_centroid_sq4(C, m)
+    ybar, b, s, sumy, ny2 = prep
+    np.testing.assert_array_equal(ybar[0], yb)
+    assert b[0] == b0 and s[0] == s0 and sumy[0] == yb.sum()
+    a, est = oracle.rbq1_assign(codes, nx2, F, popx, d, prep)
+    # direct form of Eq. final:rabitq: (1/sqrt d) sum (2 xbar_i - 1)(b + s ybar_i), fp64
+    xbar = (X - m > 0).astype(np.float64)
+    ip = ((2 * xbar - 1) * (float(b[0]) + float(s[0]) * yb)).sum(axis=1) / math.sqrt(d)
+    direct = nx2.astype(np.float64) + float(ny2[0]) - 2 * F.astype(np.float64) * ip
+    np.testing.assert_allclose(est, direct, rtol=2e-6, atol=2e-5)
+    # with sign-constant residuals and an on-grid centroid the estimate is the true distance
+    true = cdist(X.astype(np.float64), C.astype(np.float64), "sqeuclidean")[:, 0]
+    np.testing.assert_allclose(est, true, rtol=2e-6, atol=2e-5)
+
+
+def test_rbq1_hand_worked_d32_example():
+    g = json.load(open(os.path.join(GOLDEN, "rbq1_d32_hand_example.json")))
+    d = g["d"]
+    bits = np.array([(g["x_bits_word0"] >> i) & 1 for i in range(d)])
+    X = np.where(bits == 1, 1.0, -1.0).astype(np.float32)[None, :]
+    m = np.zeros(d, np.float32)
+    C = (np.arange(d) % 16).astype(np.float32)[None, :]
+    codes, nx2, F, popx = oracle.rbq1_encode(X, m)
+    assert int(codes[0, 0]) == g["x_bits_word0"]
+    assert nx2[0] == g["nx2"] and popx[0] == g["popx"]
+    assert math.isclose(float(F[0]), g["F"], rel_tol=1e-7)
+    prep = oracle.rbq1_centroid_sq4(C, m)
+    assert prep[3][0] == g["sumy"] and prep[4][0] == g["ny2"]
+    _, est = oracle.rbq1_assign(codes, nx2, F, popx, d, prep)
+    assert math.isclose(float(est[0]), g["estimate"], rel_tol=1e-6)
+    assert float(((X - C) ** 2).sum()) == g["true_l2"]
+
+
+def test_rbq1_update_is_mean_of_decoded_members():
+    r = _rng(12)
+    n, d, k = 300, 50, 5
+    X = r.standard_normal((n, d)).astype(np.float32)
+    m = oracle.rbq1_mean(X)
+    codes, nx2, F, popx = oracle.rbq1_encode(X, m)
+    e = oracle.rbq1_exponent(F)
+    mx = float(F.max())
+    assert 2.0 ** 36 < mx * 2.0 ** e <= 2.0 ** 37
+    a = r.integers(0, k - 1, n).astype(np.int32)  # cluster k-1 empty
+    C0 = r.standard_normal((k, d)).astype(np.float32)
+    C, counts = oracle.rbq1_update(codes, F, d, m, e, a, C0)
+    xbar = (X - m > 0).astype(np.float64)
+    dec = m.astype(np.float64) + F.astype(np.float64)[:, None] * (2 * xbar - 1) / math.sqrt(d)
+    for j in range(k - 1):
+        np.testing.assert_allclose(C[j], dec[a == j].mean(axis=0), rtol=1e-6, atol=1e-7)
+    np.testing.assert_array_equal(C[k - 1], C0[k - 1])
+
+
+def test_rbq1_assign_argmin_of_estimates_brute_force():
+    r = _rng(13)
+    n, d, k = 60, 40, 7
+    X = r.standard_normal((n, d)).astype(np.float32)
+    C = r.standard_normal((k, d)).astype(np.float32)
+    m = oracle.rbq1_mean(X)
+    codes, nx2, F, popx = oracle.rbq1_encode(X, m)
+    prep = oracle.rbq1_centroid_sq4(C, m)
+    a, est = oracle.rbq1_assign(codes, nx2, F, popx, d, prep)
+    ybar, b, s, sumy, ny2 = prep
+    xbar = (X - m > 0).astype(np.float64)
+    ipd = ((2 * xbar[:, None, :] - 1) * (b[None, :, None] + s[None, :, None] * ybar[None, :, :])).sum(-1) / math.sqrt(d)
+    estd = nx2[:, None] + ny2[None, :] - 2 * F[:, None] * ipd
+    top2 = np.sort(estd, axis=1)
+    clear = (top2[:, 1] - top2[:, 0]) > 1e-3 * np.abs(top2[:, 0]).max()
+    np.testing.assert_array_equal(a[clear], np.argmin(estd, axis=1)[clear])
+
+
+# ------------------------------------------------------- projection and PCA
+def test_project_matches_matmul_and_rotation_preserves_distances():
+    import synth
+
+    r = _rng(14)
+    X = r.standard_normal((40, 24)).astype(np.float32)
+    Q = synth.haar_rotation(24, 3).numpy()
+    np.testing.assert_allclose(Q.T @ Q, np.eye(24), atol=1e-12)
+    mu = X.mean(axis=0).astype(np.float32)
+    Y = oracle.project(X, Q.astype(np.float32), mu)
+    np.testing.assert_allclose(Y, (X.astype(np.float64) - mu) @ Q.astype(np.float32).astype(np.float64), rtol=1e-12, atol=1e-12)
+    np.testing.assert_allclose(cdist(Y, Y), cdist(X.astype(np.float64), X.astype(np.float64)), rtol=1e-5, atol=1e-5)
+
+
+def test_pca_recovers_axes_of_diagonal_covariance():
+    r = _rng(15)
+    lam = np.array([9.0, 4.0, 2.0, 1.0, 0.25, 0.05])
+    X = (r.standard_normal((20000, 6)) * np.sqrt(lam)).astype(np.float32)
+    mu0, cov0 = oracle.mean_cov(X)
+    np.testing.assert_allclose(cov0, np.cov(X.astype(np.float64).T, bias=True), rtol=1e-9, atol=1e-12)
+    mu, P, w = oracle.pca_fit(X, 4)
+    np.testing.assert_allclose(np.abs(P), np.eye(6)[:, :4], atol=0.03)
+    assert np.all(np.diag(P[:4, :4]) > 0)  # sign fix: largest entry positive
+    np.testing.assert_allclose(w, lam[:4], rtol=0.05)
+    # full-rank PCA is a rotation: pairwise distances are preserved
+    _, Pf, _ = oracle.pca_fit(X[:500], 6)
+    Y = oracle.project(X[:50], Pf.astype(np.float32), mu0.astype(np.float32))
+    np.testing.assert_allclose(cdist(Y, Y), cdist(X[:50].astype(np.float64), X[:50].astype(np.float64)), rtol=1e-5, atol=1e-5)
+
+
+def test_round_bf16_matches_torch_and_ties_to_even():
+    import torch
+
+    r = _rng(16)
+    f = r.standard_normal(4000).astype(np.float32)
+    want = torch.from_numpy(f).to(torch.bfloat16).view(torch.int16).numpy().view(np.uint16)
+    np.testing.assert_array_equal(oracle.round_bf16(f.astype(np.float64)), want)
+    # exact halfway cases: 1 + 2^-8 lies between 1 and 1 + 2^-7 -> even (1.0)
+    got = oracle.round_bf16(np.array([1 + 2.0 ** -8, 1 + 3 * 2.0 ** -8, 1 + 2.0 ** -8 + 2.0 ** -30]))
+    np.testing.assert_array_equal(oracle.bf16_to_f32(got), np.array([1.0, 1 + 2.0 ** -6, 1 + 2.0 ** -7], np.float32))
