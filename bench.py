@@ -1,0 +1,413 @@
+#!/usr/bin/env python
+"""Benchmark of the Lloyd k-means hot path on GB300.
+
+Workload: 1,000,000 unit-norm synthetic embeddings, d = 768 (2,000-component
+Gaussian mixture, per-dimension variance (1+j)^-0.5, Haar rotation, L2
+normalisation), k = 1,000, clustered both as raw fp32 and as RabitQ 1-bit
+codes.  One step = one Lloyd iteration (assign + update) of each
+representation, i.e. 2 * N * k point-centroid distances.  Metric:
+point-centroid distances per second per Lloyd iteration.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+
+N > 1 runs under torchrun, one rank per GPU: every rank clusters its own
+1M-point shard (weak scaling) and the update's cluster sums and counts are
+all-reduced once per representation per step (the path's one exchange).
+--impl reference times the CPU oracle on a bounded sample of the workload.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+N_POINTS, DIM, K, N_COMP = 1_000_000, 768, 1000, 2000
+METRIC = "k-means point·centroid distances/s per Lloyd iter (1 GB300); % of roofline"
+WORKLOAD = "emb1m_d768: N=1,000,000 x d=768 unit-norm GMM embeddings, k=1,000; fp32 + RabitQ 1-bit"
+SM_COUNT = 152
+# POPC results per clock per SM used for the 1-bit kernel's ALU roofline.
+POPC_PER_CLK_SM = 16
+
+
+def env_rank():
+    return (int(os.environ.get("RANK", "0")), int(os.environ.get("LOCAL_RANK", "0")),
+            int(os.environ.get("WORLD_SIZE", "1")))
+
+
+def load_peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        with open(p) as f:
+            j = json.load(f)
+        return {"hbm_gbs": j["hbm_gbs"], "bf16_tflops": j["bf16_tflops"],
+                "bf16_tflops_sustained": j.get("bf16_tflops_sustained", j["bf16_tflops"]),
+                "sm_max_mhz": j.get("sm_max_mhz", 2070.0), "source": "measured"}
+    return {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0, "sm_max_mhz": 2070.0,
+            "source": "fallback"}
+
+
+class ClockSampler:
+    """nvidia-smi samples (200 ms) of SM clock and throttle reasons while running."""
+
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index):
+        self.gpu_index = gpu_index
+        self.proc = None
+        self.lines = []
+        self.thread = None
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits", "-lms", "200",
+                 "-i", str(self.gpu_index)], stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except (OSError, ValueError):
+            self.proc = None
+            return
+        self.thread = threading.Thread(target=self._read, daemon=True)
+        self.thread.start()
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.lines.append(line.strip())
+
+    def stop(self):
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        time.sleep(0.25)
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        if self.thread:
+            self.thread.join(timeout=2)
+        sm, smax, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for ln in self.lines:
+            parts = [p.strip() for p in ln.split(",")]
+            if len(parts) < 9:
+                continue
+            try:
+                sm.append(float(parts[1]))
+                smax.append(float(parts[2]))
+            except ValueError:
+                continue
+            for nm, v in zip(names, parts[5:9]):
+                if v.lower() == "active":
+                    reasons.add(nm)
+        if not sm:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["no samples"], "samples": 0}
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(smax), "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+# ----------------------------------------------------------------------------
+def cpu_baseline_sample(X_host, C32, codes, nx2, F, popx, m, e, Cr, budget_s=12.0):
+    """Oracle (as it stands) on a bounded row sample: one Lloyd iteration of
+    each representation.  Returns (distances/s, rows, seconds, threads)."""
+    import oracle
+
+    def one(ns):
+        t0 = time.perf_counter()
+        a, _, _ = oracle.assign_f32(X_host[:ns], C32)
+        oracle.update_f32(X_host[:ns], a, C32)
+        prep = oracle.rbq1_centroid_sq4(Cr, m)
+        ar, _ = oracle.rbq1_assign(codes[:ns], nx2[:ns], F[:ns], popx[:ns], DIM, prep)
+        oracle.rbq1_update(codes[:ns], F[:ns], DIM, m, e, ar, Cr)
+        return time.perf_counter() - t0
+
+    t0 = one(500)
+    ns = int(min(X_host.shape[0], max(500, 500 * budget_s / max(t0, 1e-3))))
+    t = one(ns)
+    return 2.0 * ns * K / t, ns, t, oracle.num_threads()
+
+
+def run_ours(args):
+    import numpy as np
+    import torch
+
+    import paper_2608_14648_gb300 as skm
+    import synth
+
+    rank, local_rank, world = env_rank()
+    torch.cuda.set_device(local_rank)
+    dev = torch.device("cuda", local_rank)
+    dist = None
+    if world > 1:
+        import torch.distributed as dist
+
+        dist.init_process_group("nccl")
+    peaks = load_peaks()
+
+    # ---- inputs (per-rank shard), resident in HBM before timing -------------
+    X = synth.gmm_points(N_POINTS, DIM, N_COMP, seed=rank, device=dev)
+    idx = synth.forgy_indices(N_POINTS, K, seed=0).to(dev)
+    C32 = X[idx].clone()
+    if world > 1:
+        dist.broadcast(C32, 0)
+    pts32 = skm.Points(skm.REPR_F32, X, DIM)
+    q = skm.skm_quantize(skm.REPR_RBQ1, X)
+    if world > 1:  # global mean, then re-encode; global fixed-point exponent
+        dist.all_reduce(q["m"])
+        q["m"] /= world
+        q = skm.skm_quantize(skm.REPR_RBQ1, X, fit=False, m=q["m"])
+    e = skm.skm_rbq1_exponent(q["F"])
+    if world > 1:
+        et = torch.tensor([e], device=dev)
+        dist.all_reduce(et, op=dist.ReduceOp.MIN)
+        e = int(et.item())
+    ptsR = skm.rbq1_points(q, DIM, e)
+    Cr, _, _, _, _ = skm.skm_fit(ptsR, K, 0, init_idx=idx, want_objective=False, want_dist=False)
+    if world > 1:
+        dist.broadcast(Cr, 0)
+
+    wsA32 = skm.workspace(skm.OP_ASSIGN, pts32, K)
+    wsU32 = skm.workspace(skm.OP_UPDATE, pts32, K)
+    wsAR = skm.workspace(skm.OP_ASSIGN, ptsR, K)
+    wsUR = skm.workspace(skm.OP_UPDATE, ptsR, K)
+    a32 = torch.empty(N_POINTS, dtype=torch.int32, device=dev)
+    aR = torch.empty(N_POINTS, dtype=torch.int32, device=dev)
+    cnt32 = torch.zeros(K, dtype=torch.int64, device=dev)
+    cntR = torch.zeros(K, dtype=torch.int64, device=dev)
+    part32 = torch.zeros(K, DIM, dtype=torch.float64, device=dev) if world > 1 else None
+    partR = torch.zeros(K, DIM + 1, dtype=torch.int64, device=dev) if world > 1 else None
+    stream = torch.cuda.current_stream()
+    ev = {name: [] for name in ("a32", "aR")}
+
+    def lloyd(pts, C, a, cnt, part, wsA, wsU, key, record):
+        if record:
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record(stream)
+        skm.skm_assign(pts, C, K, want_dist=False, ws=wsA, out=a)
+        if record:
+            e1.record(stream)
+            ev[key].append((e0, e1))
+        if part is None:
+            skm.skm_update(pts, a, C, counts=cnt, ws=wsU)
+        else:
+            part.zero_()
+            cnt.zero_()
+            skm.skm_update(pts, a, None, counts=cnt, partial=part, ws=wsU)
+            dist.all_reduce(part)
+            dist.all_reduce(cnt)
+            skm.skm_update_finalize(pts, part, cnt, C)
+
+    def step(record):
+        lloyd(pts32, C32, a32, cnt32, part32, wsA32, wsU32, "a32", record)
+        lloyd(ptsR, Cr, aR, cntR, partR, wsAR, wsUR, "aR", record)
+
+    for _ in range(args.warmup):
+        step(False)
+    torch.cuda.synchronize()
+    if world > 1:
+        dist.barrier()
+    clocks = ClockSampler(local_rank)
+    clocks.start()
+    torch.cuda.synchronize()
+    launches0 = skm.skm_kernel_launches()
+    t_start, t_end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    t_start.record(stream)
+    for _ in range(args.steps):
+        step(True)
+    t_end.record(stream)
+    torch.cuda.synchronize()
+    if world > 1:
+        dist.barrier()
+    launches = skm.skm_kernel_launches() - launches0
+    clk = clocks.stop()
+    ms = t_start.elapsed_time(t_end)
+    if world > 1:
+        t = torch.tensor([ms], device=dev, dtype=torch.float64)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        ms = float(t.item())
+    ms_step = ms / args.steps
+    value = world * 2.0 * N_POINTS * K * args.steps / (ms / 1e3)
+
+    # ---- roofline of the dominant kernel --------------------------------------
+    t_a32 = statistics.mean(a.elapsed_time(b) for a, b in ev["a32"])
+    t_aR = statistics.mean(a.elapsed_time(b) for a, b in ev["aR"])
+    long_region = ms > 1000.0
+    bf16_peak = peaks["bf16_tflops_sustained"] if long_region else peaks["bf16_tflops"]
+    flops_a32 = 2.0 * N_POINTS * K * DIM
+    W = (DIM + 31) // 32
+    popc_aR = float(N_POINTS) * K * 4 * W
+    popc_peak = SM_COUNT * POPC_PER_CLK_SM * peaks["sm_max_mhz"] * 1e6  # per second
+    kernels = {
+        "assign_f32": {"ms": t_a32, "bound": "tensor", "achieved": flops_a32 / (t_a32 / 1e3) / 1e12,
+                       "peak": bf16_peak, "unit": "TFLOP/s",
+                       "algorithmic": f"2*N*k*d = {flops_a32:.3e} flop per launch"},
+        "assign_rbq1": {"ms": t_aR, "bound": "alu", "achieved": popc_aR / (t_aR / 1e3) / 1e12, "peak":
+                        popc_peak / 1e12, "unit": "Tpopc/s",
+                        "algorithmic": f"N*k*4*ceil(d/32) = {popc_aR:.3e} POPC per launch"},
+    }
+    for kd in kernels.values():
+        kd["frac"] = kd["achieved"] / kd["peak"]
+    dom = max(kernels, key=lambda n: kernels[n]["ms"])
+    kd = kernels[dom]
+    roofline = {"bound": kd["bound"], "achieved": round(kd["achieved"], 4), "peak": round(kd["peak"], 4),
+                "unit": kd["unit"], "frac": round(kd["frac"], 5), "traffic": None, "kernel": dom,
+                "peak_source": f"{peaks['source']} ({'sustained' if long_region else 'burst'} bf16)"
+                if kd["bound"] == "tensor" else f"{SM_COUNT} SMs x {POPC_PER_CLK_SM} POPC/clk x "
+                                                f"{peaks['sm_max_mhz']:.0f} MHz"}
+
+    # ---- end to end through the C ABI with host buffers ----------------------
+    e2e = None
+    if not args.no_e2e:
+        X_host = torch.empty(N_POINTS, DIM, dtype=torch.float32, pin_memory=True)
+        X_host.copy_(X)
+        C_host32 = torch.empty(K, DIM, dtype=torch.float32, pin_memory=True)
+        C_hostR = torch.empty(K, DIM, dtype=torch.float32, pin_memory=True)
+        C_host32.copy_(C32)
+        C_hostR.copy_(Cr)
+        a_host = torch.empty(2, N_POINTS, dtype=torch.int32, pin_memory=True)
+        Xd2 = torch.empty_like(X)
+        Cd32 = torch.empty_like(C32)
+        CdR = torch.empty_like(Cr)
+        pts2 = skm.Points(skm.REPR_F32, Xd2, DIM)
+        h2d = X_host.numel() * 4 + 2 * K * DIM * 4
+        d2h = 2 * N_POINTS * 4 + 2 * K * DIM * 4
+        e2e_steps = max(2, min(args.steps, 5))
+        torch.cuda.synchronize()
+        if world > 1:
+            dist.barrier()
+        s0, s1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        s0.record(stream)
+        for _ in range(e2e_steps):
+            Xd2.copy_(X_host, non_blocking=True)
+            Cd32.copy_(C_host32, non_blocking=True)
+            CdR.copy_(C_hostR, non_blocking=True)
+            qq = skm.skm_quantize(skm.REPR_RBQ1, Xd2, fit=False, m=q["m"])
+            pR2 = skm.rbq1_points(qq, DIM, e)
+            skm.skm_assign(pts2, Cd32, K, want_dist=False, ws=wsA32, out=a32)
+            skm.skm_update(pts2, a32, Cd32, counts=cnt32, ws=wsU32)
+            skm.skm_assign(pR2, CdR, K, want_dist=False, ws=wsAR, out=aR)
+            skm.skm_update(pR2, aR, CdR, counts=cntR, ws=wsUR)
+            a_host[0].copy_(a32, non_blocking=True)
+            a_host[1].copy_(aR, non_blocking=True)
+            C_host32.copy_(Cd32, non_blocking=True)
+            C_hostR.copy_(CdR, non_blocking=True)
+        s1.record(stream)
+        torch.cuda.synchronize()
+        ems = s0.elapsed_time(s1)
+        if world > 1:
+            t = torch.tensor([ems], device=dev, dtype=torch.float64)
+            dist.all_reduce(t, op=dist.ReduceOp.MAX)
+            ems = float(t.item())
+        e2e = {"value": world * 2.0 * N_POINTS * K * e2e_steps / (ems / 1e3), "unit": "distances/s",
+               "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "steps": e2e_steps,
+               "ms_per_step": ems / e2e_steps,
+               "path": "pinned host fp32 points -> H2D -> skm_quantize(RBQ1) -> skm_assign/skm_update "
+                       "(fp32, 1-bit) -> D2H assignments + centroids"}
+
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        h = {k2: v.cpu().numpy() for k2, v in q.items()}
+        codes = h["codes"].view(np.uint32)
+        X_host_np = X[:200_000].cpu().numpy()
+        v, ns, t, cores = cpu_baseline_sample(X_host_np, C32.cpu().numpy(), codes, h["nx2"], h["F"], h["popx"],
+                                              h["m"], e, Cr.cpu().numpy())
+        cpu = {"value": v, "unit": "distances/s", "cores": cores, "kind": "oracle",
+               "sample": f"{ns} of {N_POINTS} rows, one Lloyd iteration (assign + update) of fp32 and 1-bit "
+                         f"against all {K} centroids, {t:.1f} s"}
+
+    if rank == 0:
+        line = {
+            "metric": METRIC, "value": value, "unit": "distances/s", "n_gpus": world, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": ms_step, "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "f32 (bf16 screen + fp32 rescore) / u32 popcount",
+            "data": "synthetic (seeded GMM embeddings, generated on the GPU)",
+            "config": {"workload": WORKLOAD, "n": N_POINTS, "d": DIM, "k": K, "reprs": ["f32", "rbq1"],
+                       "step": "one Lloyd iteration (assign + update) per representation",
+                       "l2": "inputs larger than L2 (3.1 GB fp32 points streamed every step)",
+                       "parallelism": f"dp{world}"},
+            "roofline": roofline, "kernels": kernels, "cpu_baseline": cpu, "e2e": e2e, "clocks": clk,
+            "gpu_launches": int(launches),
+        }
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        dist.destroy_process_group()
+
+
+def run_reference(args):
+    """CPU oracle as it stands, on the host cores, on a bounded sample."""
+    import numpy as np
+
+    rank, _, world = env_rank()
+    if rank != 0:
+        return
+    import oracle
+    import synth
+
+    ns = 4000
+    X = synth.gmm_points(ns, DIM, N_COMP, seed=0).numpy()
+    idx = synth.forgy_indices(ns, K, seed=0).numpy()
+    C32 = X[idx].copy()
+    m = oracle.rbq1_mean(X)
+    codes, nx2, F, popx = oracle.rbq1_encode(X, m)
+    e = oracle.rbq1_exponent(F)
+    Cr = oracle.rbq1_decode_points(codes, F, DIM, m, e, idx)
+
+    def step(rows):
+        nonlocal C32, Cr
+        a, _, _ = oracle.assign_f32(X[:rows], C32)
+        C32, _ = oracle.update_f32(X[:rows], a, C32)
+        prep = oracle.rbq1_centroid_sq4(Cr, m)
+        ar, _ = oracle.rbq1_assign(codes[:rows], nx2[:rows], F[:rows], popx[:rows], DIM, prep)
+        Cr, _ = oracle.rbq1_update(codes[:rows], F[:rows], DIM, m, e, ar, Cr)
+
+    t0 = time.perf_counter()
+    step(500)
+    t1 = time.perf_counter() - t0
+    budget = 150.0 / max(1, args.steps + args.warmup)
+    rows = int(min(ns, max(500, 500 * budget / max(t1, 1e-3))))
+    for _ in range(args.warmup):
+        step(rows)
+    t0 = time.perf_counter()
+    for _ in range(args.steps):
+        step(rows)
+    t = time.perf_counter() - t0
+    value = 2.0 * rows * K * args.steps / t
+    sample = f"{rows} rows of the {WORKLOAD} recipe, one Lloyd iteration per representation per step"
+    line = {"impl": "reference", "metric": METRIC, "value": value, "unit": "distances/s", "n_gpus": world,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * t / args.steps,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64 (oracle)",
+            "data": "synthetic (seeded GMM embeddings)",
+            "config": {"workload": WORKLOAD, "n": N_POINTS, "d": DIM, "k": K, "reprs": ["f32", "rbq1"],
+                       "parallelism": "host cores"},
+            "cpu_baseline": {"value": value, "unit": "distances/s", "kind": "oracle", "cores": oracle.num_threads(),
+                             "sample": sample},
+            "e2e": {"value": value, "unit": "distances/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=10)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args()
+    if args.warmup < 3:
+        print("warning: fewer than 3 warm-up steps", file=sys.stderr)
+    if args.impl == "reference":
+        run_reference(args)
+    else:
+        run_ours(args)
+
+
+if __name__ == "__main__":
+    main()

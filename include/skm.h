@@ -1,0 +1,258 @@
+/*
+ * skm.h -- C ABI of libskm, the GB300 (sm_103a) Lloyd k-means hot path for
+ * clustering embeddings after dimensionality reduction, quantization or with
+ * dimension pruning ("Stop Indexing at Full Precision: Revisiting Clustering
+ * for Vector Embeddings", arxiv 2608.14648).
+ *
+ * Conventions shared by every entry point
+ * ---------------------------------------
+ *  - Data pointers are DEVICE pointers owned by the caller, row-major and
+ *    contiguous, unless an argument says "host".  The library never frees or
+ *    retains a caller pointer after the call returns.
+ *  - `stream` is a cudaStream_t passed as void* (NULL = the legacy default
+ *    stream).  Calls are asynchronous on that stream unless documented
+ *    otherwise; outputs are valid once the stream has reached the call.
+ *  - Scratch memory: entry points that need it take `ws`/`ws_bytes`, a device
+ *    buffer of at least skm_workspace_size(...) bytes, 256-byte aligned,
+ *    owned by the caller and not used by anything else on other streams while
+ *    the call's work is in flight.  The library itself never allocates device
+ *    memory.
+ *  - Return value: SKM_OK (0) or an skm_status error code.  Arguments are
+ *    validated on the host BEFORE any launch; on an error nothing has been
+ *    enqueued and outputs are untouched.  skm_last_error() returns a
+ *    thread-local description of the last error.  No C++ exception crosses
+ *    the ABI.
+ *  - Distances are squared L2.  Ties in every argmin go to the LOWEST
+ *    centroid index.
+ *  - Limits: 1 <= d <= 4096, 1 <= k <= 65536, 1 <= n < 2^31 (RBQ1: n <= 2^24).
+ */
+#ifndef SKM_H
+#define SKM_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* ---- status codes ------------------------------------------------------ */
+typedef enum skm_status {
+    SKM_OK = 0,
+    SKM_ERR_INVALID_ARG = 1,  /* bad shape, null pointer, k > n, bad enum    */
+    SKM_ERR_UNSUPPORTED = 2,  /* valid but outside this build's limits       */
+    SKM_ERR_CUDA = 3,         /* a CUDA runtime/driver call failed            */
+    SKM_ERR_NO_MEMORY = 4,    /* ws_bytes smaller than skm_workspace_size()  */
+    SKM_ERR_TIMEOUT = 5,      /* a bounded device wait gave up               */
+    SKM_ERR_DEVICE_CHECK = 6  /* a device-side check recorded a failure      */
+} skm_status;
+
+/* ---- representations of the points being clustered (Table 1) ---------- */
+typedef enum skm_repr {
+    SKM_REPR_F32 = 0,  /* float32 [n][d]                                    */
+    SKM_REPR_SQ8 = 1,  /* uint8 SQ8 codes [n][d] (Section 3.1, per-dim b,s)  */
+    SKM_REPR_RBQ1 = 2, /* RabitQ 1-bit codes uint32 [n][ceil(d/32)]
+                          (bit j of word w = dimension 32w+j) + factors     */
+    SKM_REPR_BF16 = 3  /* bfloat16 bit patterns uint16 [n][d] (projected
+                          points stored in bf16), fp32 centroids            */
+} skm_repr;
+
+typedef enum skm_dtype { SKM_DTYPE_F32 = 0, SKM_DTYPE_BF16 = 1 } skm_dtype;
+
+/* Points being clustered.  Which fields are read depends on repr. */
+typedef struct skm_data {
+    int32_t repr;       /* skm_repr                                          */
+    int32_t d;          /* dimensions                                        */
+    int64_t n;          /* points                                            */
+    const void *x;      /* the points / codes, layout per repr               */
+    /* RBQ1 only (outputs of skm_quantize): per-point factors of Eq. rabitq_l2 */
+    const float *nx2;   /* ||x_r - m||^2                 [n]                 */
+    const float *F;     /* ||x_r - m|| / <xbar, x>       [n]                 */
+    const int32_t *popx;/* number of set bits            [n]                 */
+    const float *m;     /* centring mean m               [d]                 */
+    int32_t rbq1_exp;   /* fixed-point exponent e of the decode-average
+                           (skm_rbq1_exponent); fit() computes it itself     */
+    int32_t reserved0;
+} skm_data;
+
+/* Optional per-call statistics (host struct, filled after the call's work
+ * completes only when the call synchronises, i.e. skm_fit). */
+typedef struct skm_stats {
+    int64_t rescored_rows;    /* F32/BF16: rows whose screen was not decisive */
+    int64_t fallback_rows;    /* F32/BF16: rows rescanned over all k in fp32  */
+    int64_t empty_clusters;   /* after the last update                         */
+    int64_t reserved[5];
+} skm_stats;
+
+const char *skm_last_error(void);
+int skm_version(void); /* major*10000 + minor*100 + patch */
+
+/* Number of CUDA kernels this library has enqueued in this process so far
+ * (host-side counter over all threads and devices; diagnostic only, e.g. to
+ * count the kernels inside a timed region). */
+uint64_t skm_kernel_launches(void);
+
+/* Bytes of scratch needed by op for these points and k centroids.
+ * op: 0 = skm_assign, 1 = skm_update, 2 = skm_fit, 3 = skm_quantize,
+ *     4 = skm_pca_fit.
+ * Returns 0 with skm_last_error() set when the arguments are invalid. */
+size_t skm_workspace_size(int op, const skm_data *x, int k);
+
+/* ------------------------------------------------------------------------
+ * Projection (Section 3.1: JLT / PCA; the random orthogonal rotation that
+ * SuperKMeans and RabitQ require).  Y = (X - mean) P.
+ *   X      float32 [n][d]
+ *   mean   float32 [d] or NULL (no centring)
+ *   P      float32 [d][d_out], row-major (column j = output direction j)
+ *   Y      out_dtype [n][d_out]: SKM_DTYPE_F32 (float) or SKM_DTYPE_BF16
+ *          (bf16 bit patterns, rounded half to even from the fp32 result)
+ * fp32 arithmetic.  d_out <= d.
+ * ------------------------------------------------------------------------ */
+int skm_project(const float *X, int64_t n, int d, const float *mean, const float *P,
+                int d_out, int out_dtype, void *Y, void *stream);
+
+/* Haar-random orthogonal d x d matrix (HOST helper, host output P_host[d][d],
+ * float32 row-major): Householder QR of a Gaussian matrix drawn with
+ * Philox4x32-10 + Box-Muller from `seed`, signs fixed so R has a positive
+ * diagonal.  Synchronous, no GPU use. */
+int skm_make_rotation(uint64_t seed, int d, float *P_host);
+
+/* PCA fit (Section 3.1 "PCA"): mean and population covariance of X on the
+ * GPU (fp32 products, fp64 accumulation), then a symmetric eigen-
+ * decomposition on the host (fp64 Householder tridiagonalisation + implicit
+ * QL).  Outputs (device): mean float32[d]; P float32 [d][d_out] whose columns
+ * are the top-d_out eigenvectors by descending eigenvalue, each signed so its
+ * largest-magnitude entry is positive; eigvals float32[d_out] (may be NULL).
+ * Synchronises `stream` (the covariance is copied to the host). */
+int skm_pca_fit(const float *X, int64_t n, int d, int d_out, float *mean, float *P,
+                float *eigvals, void *ws, size_t ws_bytes, void *stream);
+
+/* ------------------------------------------------------------------------
+ * Quantization of the points before clustering (Section 3.1).
+ *  repr = SKM_REPR_SQ8: per-dimension bias b_i = min over points and scale
+ *    s_i = (max - b_i) / 255 (s_i = 1 for a flat dimension) when fit != 0,
+ *    else the supplied b, s are used; code = clip(round((x - b)/s), 0, 255)
+ *    in fp32, rounding half to even.  Outputs: codes uint8[n][d], b,s [d].
+ *  repr = SKM_REPR_RBQ1 (RabitQ, 1-bit): mean m (fp64 sum, rounded to fp32)
+ *    when fit != 0, else the supplied m; r = x - m; bit i = (r_i > 0);
+ *    nx2 = ||r||^2; F = sqrt(d) ||r||^2 / ||r||_1 (0 when r = 0), i.e.
+ *    ||r|| / <xbar, x>; popx = set bits.  Outputs: codes uint32[n][W],
+ *    W = ceil(d/32), bit j of word w = dim 32w+j (unused high bits are 0);
+ *    nx2, F float[n]; popx int32[n]; m float[d].
+ *  X float32 [n][d].  The x rows are assumed already rotated when RabitQ's
+ *  random rotation is wanted (skm_project with skm_make_rotation's P).
+ * ------------------------------------------------------------------------ */
+typedef struct skm_quant_params {
+    int32_t fit;   /* 1: fit b,s (SQ8) or m (RBQ1) from X; 0: use supplied  */
+    int32_t reserved0;
+    float *b;      /* SQ8 bias  [d] (device; output when fit, else input)    */
+    float *s;      /* SQ8 scale [d]                                          */
+    float *m;      /* RBQ1 mean [d]                                          */
+    float *nx2;    /* RBQ1 outputs [n]                                       */
+    float *F;
+    int32_t *popx;
+} skm_quant_params;
+
+int skm_quantize(int repr, const float *X, int64_t n, int d, skm_quant_params *qp,
+                 void *codes, void *ws, size_t ws_bytes, void *stream);
+
+/* Fixed-point exponent e of the RBQ1 decode-average: e = 37 - ceil(log2 max F)
+ * (0 when every F is 0), so round(F 2^e) <= 2^37 and the per-cluster sums of
+ * up to 2^24 points are exact in int64.  Writes *e_host; synchronises. */
+int skm_rbq1_exponent(const float *F, int64_t n, int *e_host, void *ws, size_t ws_bytes,
+                      void *stream);
+
+/* ------------------------------------------------------------------------
+ * Assignment, Section 2.3 STEP 2: assign[p] = argmin_j dist(x_p, c_j).
+ *  C (device), per repr:
+ *   F32  float [k][d] centroids.  Exact fp32 nearest centroid: a bf16
+ *        tensor-core screen with a rigorous per-pair error bound, fp32
+ *        rescoring (direct differences) of every centroid the bound cannot
+ *        rule out, and an fp32 scan over all k for rows the screen could not
+ *        narrow down.  dist = fp32 sum of squared differences.
+ *   BF16 float [k][d] centroids against bf16 points; exact dimension
+ *        pruning over 32-dimension prefix blocks (a centroid is dropped as
+ *        soon as its partial distance exceeds the row's current best).
+ *   SQ8  uint8 [k][d] centroid codes; exact integer code-space distance
+ *        sum (xbar_i - cbar_i)^2 (dist is that integer, as float).
+ *   RBQ1 float [k][d] decoded centroids; per iteration each centroid is
+ *        re-encoded with per-centroid SQ4 (b = min, s = (max-b)/15 of
+ *        c - m) and the distance is the estimator of Eq. rabitq_l2 with
+ *        Eq. final:rabitq, evaluated in fp32 in the order
+ *          t1 = s (2P - sum ybar), t2 = b (2 popx - d),
+ *          ip = (t1 + t2) * fl(1/sqrt d), dist = (nx2 + ny2) - 2 (F ip)
+ *        where P = sum_i xbar_i ybar_i is an exact AND+popcount sum.
+ *  assign int32[n] (required); dist float[n] (may be NULL).
+ *  prev_assign int32[n] or NULL: BF16 only, seeds the pruning bound with
+ *  the distance to the previous centroid (results do not depend on it).
+ * ------------------------------------------------------------------------ */
+int skm_assign(const skm_data *x, const void *C, int k, const int32_t *prev_assign,
+               int32_t *assign, float *dist, void *ws, size_t ws_bytes, void *stream);
+
+/* ------------------------------------------------------------------------
+ * Update, Section 2.3 STEP 3 (and the quantized-domain variants of 3.1).
+ *  C_inout (device), per repr as in skm_assign; clusters with no member keep
+ *  their centroid.  counts int64[k] (device, output).
+ *   F32/BF16  c_j = mean of members (fp32 sums per cluster)
+ *   SQ8       cbar_j = round-half-even(sum of member codes / count), exact
+ *   RBQ1      fused decode-average: c_ji = m_i + ((2 T_ji - U_j) 2^-e
+ *             / count_j) / sqrt(d) in fp64, rounded to fp32, where
+ *             T_ji = sum Fq xbar_i, U_j = sum Fq, Fq = round(F 2^e) (int64,
+ *             exact), e = x->rbq1_exp.
+ *  partial != NULL selects the sharded form: nothing is finalised; the
+ *  cluster sums are ADDED into `partial` and the member counts into
+ *  `counts` (both zeroed by the caller before the first shard) so that
+ *  shards can be merged (skm_merge_partials) and finalised
+ *  (skm_update_finalize).  partial layout: F32/BF16 double[k][d];
+ *  SQ8 int64[k][d]; RBQ1 int64[k][d+1] (T then U).
+ * ------------------------------------------------------------------------ */
+int skm_update(const skm_data *x, const int32_t *assign, int k, void *C_inout,
+               int64_t *counts, void *partial, void *ws, size_t ws_bytes, void *stream);
+
+/* dst += src over `count` elements of the partial layout (elem_type 0 =
+ * double, 1 = int64); device pointers. */
+int skm_merge_partials(void *dst, const void *src, int64_t count, int elem_type, void *stream);
+
+/* Finalise merged partial sums into centroids (same rules as skm_update). */
+int skm_update_finalize(const skm_data *x, const void *partial, const int64_t *counts,
+                        int k, void *C_inout, void *stream);
+
+/* ------------------------------------------------------------------------
+ * Lloyd k-means, Section 2.3: `iters` x (STEP 2 assign, STEP 3 update), then
+ * STEP 2 once more for the final assignment.
+ *  cfg->iters >= 0.  Initial centroids: C_init (device, per-repr layout of
+ *  skm_assign) when non-NULL, else the points init_idx[0..k) (device int64,
+ *  Forgy, STEP 1): F32/BF16 rows, SQ8 codes, RBQ1 decoded points (the
+ *  decode-average of one member).
+ *  Outputs (device): C_out (per-repr layout), assign_out int32[n],
+ *  dist_out float[n] or NULL (from the final assignment).
+ *  objective_host (host, iters+1 doubles, may be NULL): sum of the
+ *  assignment's dist at each STEP 2 (fp64 sum of the per-row values).
+ *  stats_host may be NULL.  Synchronises `stream` before returning.
+ * ------------------------------------------------------------------------ */
+typedef struct skm_fit_config {
+    int32_t k;
+    int32_t iters;
+    int32_t reserved[6];
+} skm_fit_config;
+
+int skm_fit(const skm_fit_config *cfg, const skm_data *x, const void *C_init,
+            const int64_t *init_idx, void *C_out, int32_t *assign_out, float *dist_out,
+            double *objective_host, skm_stats *stats_host, void *ws, size_t ws_bytes,
+            void *stream);
+
+/* Objective helpers (reporting, Section 4 WCSS): fp64 sum over n of
+ * ||x_p - c_{a_p}||^2 with x float32 [n][d] (or bf16 bits when x_is_bf16)
+ * and C float32 [k][d].  Writes *out_host; synchronises. */
+int skm_objective(const void *X, int x_is_bf16, int64_t n, int d, const float *C, int k,
+                  const int32_t *assign, double *out_host, void *ws, size_t ws_bytes,
+                  void *stream);
+
+/* SQ8 reconstruction x ~ code * s + b (fp32): codes uint8[n][d] -> Y float[n][d]. */
+int skm_sq8_decode(const uint8_t *codes, int64_t n, int d, const float *b, const float *s,
+                   float *Y, void *stream);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* SKM_H */

@@ -1,0 +1,315 @@
+"""Python binding of libskm, the GB300 Lloyd k-means hot path (C ABI in
+include/skm.h).
+
+Argument marshalling only: torch tensors provide device memory and streams,
+every step of the path runs in the CUDA kernels of libskm.so.  There is no
+fallback: if the library is missing, importing the binding's entry points
+raises.  Function names match the C entry points.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+
+import torch
+
+__all__ = [
+    "REPR_F32", "REPR_SQ8", "REPR_RBQ1", "REPR_BF16", "SkmError", "lib", "lib_path", "Data",
+    "skm_version", "skm_kernel_launches", "skm_workspace_size", "skm_project", "skm_make_rotation", "skm_pca_fit",
+    "skm_quantize", "skm_rbq1_exponent", "skm_assign", "skm_update", "skm_merge_partials",
+    "skm_update_finalize", "skm_fit", "skm_objective", "skm_sq8_decode", "EXPORTED_SYMBOLS",
+]
+
+REPR_F32, REPR_SQ8, REPR_RBQ1, REPR_BF16 = 0, 1, 2, 3
+DTYPE_F32, DTYPE_BF16 = 0, 1
+OP_ASSIGN, OP_UPDATE, OP_FIT, OP_QUANTIZE, OP_PCA = 0, 1, 2, 3, 4
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+_LIB_PATH = os.path.join(_HERE, "_build", "libskm.so")
+_lib = None
+
+# Every entry point declared in include/skm.h.
+EXPORTED_SYMBOLS = [
+    "skm_last_error", "skm_version", "skm_kernel_launches", "skm_workspace_size", "skm_project", "skm_make_rotation",
+    "skm_pca_fit", "skm_quantize", "skm_rbq1_exponent", "skm_assign", "skm_update",
+    "skm_merge_partials", "skm_update_finalize", "skm_fit", "skm_objective", "skm_sq8_decode",
+]
+
+
+class SkmError(RuntimeError):
+    def __init__(self, code, msg):
+        super().__init__(f"libskm error {code}: {msg}")
+        self.code = code
+
+
+class Data(ctypes.Structure):
+    """skm_data (include/skm.h)."""
+
+    _fields_ = [
+        ("repr", ctypes.c_int32), ("d", ctypes.c_int32), ("n", ctypes.c_int64),
+        ("x", ctypes.c_void_p), ("nx2", ctypes.c_void_p), ("F", ctypes.c_void_p),
+        ("popx", ctypes.c_void_p), ("m", ctypes.c_void_p), ("rbq1_exp", ctypes.c_int32),
+        ("reserved0", ctypes.c_int32),
+    ]
+
+
+class QuantParams(ctypes.Structure):
+    _fields_ = [
+        ("fit", ctypes.c_int32), ("reserved0", ctypes.c_int32), ("b", ctypes.c_void_p),
+        ("s", ctypes.c_void_p), ("m", ctypes.c_void_p), ("nx2", ctypes.c_void_p),
+        ("F", ctypes.c_void_p), ("popx", ctypes.c_void_p),
+    ]
+
+
+class Stats(ctypes.Structure):
+    _fields_ = [("rescored_rows", ctypes.c_int64), ("fallback_rows", ctypes.c_int64),
+                ("empty_clusters", ctypes.c_int64), ("reserved", ctypes.c_int64 * 5)]
+
+
+class FitConfig(ctypes.Structure):
+    _fields_ = [("k", ctypes.c_int32), ("iters", ctypes.c_int32), ("reserved", ctypes.c_int32 * 6)]
+
+
+def lib_path() -> str:
+    return _LIB_PATH
+
+
+def lib():
+    """The loaded libskm.so; raises if it has not been built."""
+    global _lib
+    if _lib is None:
+        if not os.path.exists(_LIB_PATH):
+            raise ImportError(f"libskm.so not found at {_LIB_PATH}: run `python -c 'import __graft_entry__ as g; g.build()'`")
+        L = ctypes.CDLL(_LIB_PATH)
+        vp, i32, i64, u64, sz = ctypes.c_void_p, ctypes.c_int, ctypes.c_int64, ctypes.c_uint64, ctypes.c_size_t
+        sig = {
+            "skm_last_error": ([], ctypes.c_char_p),
+            "skm_version": ([], i32),
+            "skm_kernel_launches": ([], ctypes.c_uint64),
+            "skm_workspace_size": ([i32, vp, i32], sz),
+            "skm_project": ([vp, i64, i32, vp, vp, i32, i32, vp, vp], i32),
+            "skm_make_rotation": ([u64, i32, vp], i32),
+            "skm_pca_fit": ([vp, i64, i32, i32, vp, vp, vp, vp, sz, vp], i32),
+            "skm_quantize": ([i32, vp, i64, i32, vp, vp, vp, sz, vp], i32),
+            "skm_rbq1_exponent": ([vp, i64, vp, vp, sz, vp], i32),
+            "skm_assign": ([vp, vp, i32, vp, vp, vp, vp, sz, vp], i32),
+            "skm_update": ([vp, vp, i32, vp, vp, vp, vp, sz, vp], i32),
+            "skm_merge_partials": ([vp, vp, i64, i32, vp], i32),
+            "skm_update_finalize": ([vp, vp, vp, i32, vp, vp], i32),
+            "skm_fit": ([vp, vp, vp, vp, vp, vp, vp, vp, vp, vp, sz, vp], i32),
+            "skm_objective": ([vp, i32, i64, i32, vp, i32, vp, vp, vp, sz, vp], i32),
+            "skm_sq8_decode": ([vp, i64, i32, vp, vp, vp, vp], i32),
+        }
+        for name, (args, res) in sig.items():
+            fn = getattr(L, name)
+            fn.argtypes = args
+            fn.restype = res
+        _lib = L
+    return _lib
+
+
+def _check(rc):
+    if rc != 0:
+        raise SkmError(rc, lib().skm_last_error().decode())
+
+
+def _ptr(t):
+    return None if t is None else ctypes.c_void_p(t.data_ptr())
+
+
+def _stream(stream=None):
+    s = stream if stream is not None else torch.cuda.current_stream()
+    return ctypes.c_void_p(s.cuda_stream)
+
+
+def _ws(nbytes, device):
+    nbytes = max(int(nbytes), 256)
+    # 256-byte alignment: the caching allocator returns 512-byte aligned blocks
+    return torch.empty(nbytes, dtype=torch.uint8, device=device)
+
+
+def _dev(t):
+    return t.device if t is not None else torch.device("cuda")
+
+
+class Points:
+    """Keeps the tensors of one skm_data alive; `.ref` is the ctypes struct."""
+
+    def __init__(self, repr_, x, d, nx2=None, F=None, popx=None, m=None, rbq1_exp=0):
+        assert x.is_contiguous()
+        self.repr, self.x, self.d = repr_, x, int(d)
+        self.nx2, self.F, self.popx, self.m = nx2, F, popx, m
+        self.n = x.shape[0]
+        self.rbq1_exp = int(rbq1_exp)
+        self.ref = Data(repr_, self.d, self.n, x.data_ptr(), _ptr(nx2), _ptr(F), _ptr(popx), _ptr(m),
+                        self.rbq1_exp, 0)
+
+    @property
+    def device(self):
+        return self.x.device
+
+
+def skm_version() -> int:
+    return lib().skm_version()
+
+
+def skm_kernel_launches() -> int:
+    return int(lib().skm_kernel_launches())
+
+
+def skm_workspace_size(op, pts: Points, k) -> int:
+    n = lib().skm_workspace_size(op, ctypes.byref(pts.ref), int(k))
+    if n == 0:
+        raise SkmError(1, lib().skm_last_error().decode())
+    return n
+
+
+def skm_project(X, P, mean=None, out_dtype=DTYPE_F32, stream=None):
+    n, d = X.shape
+    d_out = P.shape[1]
+    Y = torch.empty(n, d_out, device=X.device, dtype=torch.float32 if out_dtype == DTYPE_F32 else torch.bfloat16)
+    _check(lib().skm_project(_ptr(X), n, d, _ptr(mean), _ptr(P), d_out, out_dtype, _ptr(Y), _stream(stream)))
+    return Y
+
+
+def skm_make_rotation(seed, d):
+    out = torch.empty(d, d, dtype=torch.float32)
+    _check(lib().skm_make_rotation(int(seed), int(d), ctypes.c_void_p(out.data_ptr())))
+    return out
+
+
+def skm_pca_fit(X, d_out, stream=None):
+    n, d = X.shape
+    dummy = Points(REPR_F32, X, d)
+    ws = _ws(skm_workspace_size(OP_PCA, dummy, 1), X.device)
+    mean = torch.empty(d, device=X.device, dtype=torch.float32)
+    P = torch.empty(d, d_out, device=X.device, dtype=torch.float32)
+    w = torch.empty(d_out, device=X.device, dtype=torch.float32)
+    _check(lib().skm_pca_fit(_ptr(X), n, d, d_out, _ptr(mean), _ptr(P), _ptr(w), _ptr(ws), ws.numel(),
+                             _stream(stream)))
+    return mean, P, w
+
+
+def skm_quantize(repr_, X, fit=True, b=None, s=None, m=None, stream=None):
+    """SQ8 -> dict(codes, b, s); RBQ1 -> dict(codes, m, nx2, F, popx)."""
+    n, d = X.shape
+    dev = X.device
+    dummy = Points(REPR_F32, X, d)
+    ws = _ws(skm_workspace_size(OP_QUANTIZE, dummy, 1), dev)
+    if repr_ == REPR_SQ8:
+        b = b if b is not None else torch.empty(d, device=dev, dtype=torch.float32)
+        s = s if s is not None else torch.empty(d, device=dev, dtype=torch.float32)
+        codes = torch.empty(n, d, device=dev, dtype=torch.uint8)
+        qp = QuantParams(int(fit), 0, b.data_ptr(), s.data_ptr(), None, None, None, None)
+        _check(lib().skm_quantize(repr_, _ptr(X), n, d, ctypes.byref(qp), _ptr(codes), _ptr(ws), ws.numel(),
+                                  _stream(stream)))
+        return {"codes": codes, "b": b, "s": s}
+    if repr_ == REPR_RBQ1:
+        W = (d + 31) // 32
+        m = m if m is not None else torch.empty(d, device=dev, dtype=torch.float32)
+        codes = torch.empty(n, W, device=dev, dtype=torch.int32)
+        nx2 = torch.empty(n, device=dev, dtype=torch.float32)
+        F = torch.empty(n, device=dev, dtype=torch.float32)
+        popx = torch.empty(n, device=dev, dtype=torch.int32)
+        qp = QuantParams(int(fit), 0, None, None, m.data_ptr(), nx2.data_ptr(), F.data_ptr(), popx.data_ptr())
+        _check(lib().skm_quantize(repr_, _ptr(X), n, d, ctypes.byref(qp), _ptr(codes), _ptr(ws), ws.numel(),
+                                  _stream(stream)))
+        return {"codes": codes, "m": m, "nx2": nx2, "F": F, "popx": popx}
+    raise ValueError("repr must be REPR_SQ8 or REPR_RBQ1")
+
+
+def skm_rbq1_exponent(F, stream=None):
+    ws = _ws(1024, F.device)
+    e = ctypes.c_int(0)
+    _check(lib().skm_rbq1_exponent(_ptr(F), F.numel(), ctypes.byref(e), _ptr(ws), ws.numel(), _stream(stream)))
+    return e.value
+
+
+def workspace(op, pts: Points, k):
+    """A device workspace tensor sized for op (OP_ASSIGN, OP_UPDATE, OP_FIT)."""
+    return _ws(skm_workspace_size(op, pts, k), pts.device)
+
+
+def rbq1_points(q, d, e=None):
+    """Points for the RBQ1 representation from skm_quantize's outputs."""
+    if e is None:
+        e = skm_rbq1_exponent(q["F"])
+    return Points(REPR_RBQ1, q["codes"], d, q["nx2"], q["F"], q["popx"], q["m"], e)
+
+
+def skm_assign(pts: Points, C, k=None, prev_assign=None, want_dist=True, ws=None, stream=None, out=None,
+               dist_out=None):
+    k = C.shape[0] if k is None else k
+    dev = pts.device
+    if ws is None:
+        ws = _ws(skm_workspace_size(OP_ASSIGN, pts, k), dev)
+    assign = out if out is not None else torch.empty(pts.n, device=dev, dtype=torch.int32)
+    dist = None
+    if want_dist:
+        dist = dist_out if dist_out is not None else torch.empty(pts.n, device=dev, dtype=torch.float32)
+    _check(lib().skm_assign(ctypes.byref(pts.ref), _ptr(C), int(k), _ptr(prev_assign), _ptr(assign), _ptr(dist),
+                            _ptr(ws), ws.numel(), _stream(stream)))
+    return assign, dist
+
+
+def skm_update(pts: Points, assign, C_inout, counts=None, partial=None, ws=None, stream=None):
+    k = C_inout.shape[0] if C_inout is not None else counts.shape[0]
+    dev = pts.device
+    if ws is None:
+        ws = _ws(skm_workspace_size(OP_UPDATE, pts, k), dev)
+    if counts is None:
+        counts = torch.zeros(k, device=dev, dtype=torch.int64)
+    _check(lib().skm_update(ctypes.byref(pts.ref), _ptr(assign), int(k), _ptr(C_inout), _ptr(counts), _ptr(partial),
+                            _ptr(ws), ws.numel(), _stream(stream)))
+    return C_inout, counts
+
+
+def skm_merge_partials(dst, src, stream=None):
+    et = 0 if dst.dtype == torch.float64 else 1
+    _check(lib().skm_merge_partials(_ptr(dst), _ptr(src), dst.numel(), et, _stream(stream)))
+    return dst
+
+
+def skm_update_finalize(pts: Points, partial, counts, C_inout, stream=None):
+    _check(lib().skm_update_finalize(ctypes.byref(pts.ref), _ptr(partial), _ptr(counts), C_inout.shape[0],
+                                     _ptr(C_inout), _stream(stream)))
+    return C_inout
+
+
+def skm_fit(pts: Points, k, iters, C_init=None, init_idx=None, want_objective=True, want_dist=True,
+            ws=None, stream=None):
+    """Returns (C, assign, dist or None, objective list or None, stats dict)."""
+    dev = pts.device
+    if ws is None:
+        ws = _ws(skm_workspace_size(OP_FIT, pts, k), dev)
+    if pts.repr == REPR_SQ8:
+        C = torch.empty(k, pts.d, device=dev, dtype=torch.uint8)
+    else:
+        C = torch.empty(k, pts.d, device=dev, dtype=torch.float32)
+    assign = torch.empty(pts.n, device=dev, dtype=torch.int32)
+    dist = torch.empty(pts.n, device=dev, dtype=torch.float32) if want_dist else None
+    obj = (ctypes.c_double * (iters + 1))() if want_objective else None
+    st = Stats()
+    cfg = FitConfig(int(k), int(iters))
+    _check(lib().skm_fit(ctypes.byref(cfg), ctypes.byref(pts.ref), _ptr(C_init), _ptr(init_idx), _ptr(C),
+                         _ptr(assign), _ptr(dist), obj, ctypes.byref(st), _ptr(ws), ws.numel(), _stream(stream)))
+    stats = {"rescored_rows": st.rescored_rows, "fallback_rows": st.fallback_rows,
+             "empty_clusters": st.empty_clusters}
+    return C, assign, dist, (list(obj) if obj is not None else None), stats
+
+
+def skm_objective(X, C, assign, stream=None):
+    n, d = X.shape
+    is_bf16 = 1 if X.dtype in (torch.bfloat16, torch.int16, torch.uint16) else 0
+    ws = _ws(8192, X.device)
+    out = ctypes.c_double(0.0)
+    _check(lib().skm_objective(_ptr(X), is_bf16, n, d, _ptr(C), C.shape[0], _ptr(assign), ctypes.byref(out),
+                               _ptr(ws), ws.numel(), _stream(stream)))
+    return out.value
+
+
+def skm_sq8_decode(codes, b, s, stream=None):
+    n, d = codes.shape
+    Y = torch.empty(n, d, device=codes.device, dtype=torch.float32)
+    _check(lib().skm_sq8_decode(_ptr(codes), n, d, _ptr(b), _ptr(s), _ptr(Y), _stream(stream)))
+    return Y

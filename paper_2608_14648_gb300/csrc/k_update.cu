@@ -1,0 +1,362 @@
+// Centroid update, Section 2.3 STEP 3 (and the quantized-domain forms of
+// Section 3.1): a sort-by-cluster segmented reduction.
+//   1. histogram of assignments (shared-memory privatised counters),
+//   2. exclusive scan -> per-cluster offsets,
+//   3. scatter point ids into cluster-contiguous order,
+//   4. one CTA per cluster sums its members' rows (coalesced row reads) and
+//      finalises the centroid (or adds into caller partial sums).
+// Integer representations accumulate in int64 and are exact, so their result
+// does not depend on the member order produced by the scatter.
+#include "skm_internal.cuh"
+
+namespace skm {
+
+// ---------------------------------------------------------------- histogram
+__global__ void histogram_kernel(const int32_t *__restrict__ assign, int64_t n, int k,
+                                 int32_t *__restrict__ counts, int use_smem) {
+    extern __shared__ int32_t sh[];
+    if (use_smem) {
+        for (int j = threadIdx.x; j < k; j += blockDim.x) sh[j] = 0;
+        __syncthreads();
+    }
+    for (int64_t t = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; t < n;
+         t += (int64_t)gridDim.x * blockDim.x) {
+        const int a = assign[t];
+        if (a < 0 || a >= k) continue;  // out-of-range assignments are skipped
+        if (use_smem)
+            atomicAdd(&sh[a], 1);
+        else
+            atomicAdd(&counts[a], 1);
+    }
+    if (use_smem) {
+        __syncthreads();
+        for (int j = threadIdx.x; j < k; j += blockDim.x)
+            if (sh[j]) atomicAdd(&counts[j], sh[j]);
+    }
+}
+
+cudaError_t launch_histogram(const int32_t *assign, int64_t n, int k, int32_t *counts32,
+                             cudaStream_t st) {
+    cudaError_t e = cudaMemsetAsync(counts32, 0, sizeof(int32_t) * (size_t)k, st);
+    if (e != cudaSuccess) return e;
+    if (n == 0) return cudaSuccess;
+    const int use_smem = k <= 12288;
+    const size_t smem = use_smem ? sizeof(int32_t) * (size_t)k : 0;
+    int64_t blocks = (n + 1023) / 1024;
+    if (blocks > 152 * 4) blocks = 152 * 4;
+    histogram_kernel<<<(unsigned)blocks, 512, smem, st>>>(assign, n, k, counts32, use_smem);
+    return launched();
+}
+
+// --------------------------------------------------------------------- scan
+// Single block; each thread scans a contiguous run of counts.
+__global__ void scan_offsets_kernel(const int32_t *__restrict__ counts, int k,
+                                    int64_t *__restrict__ offsets, int64_t *__restrict__ counts64,
+                                    int accumulate) {
+    __shared__ int64_t part[1024];
+    const int t = threadIdx.x;
+    const int per = (k + blockDim.x - 1) / blockDim.x;
+    const int lo = min(k, t * per), hi = min(k, lo + per);
+    int64_t s = 0;
+    for (int j = lo; j < hi; ++j) s += counts[j];
+    part[t] = s;
+    __syncthreads();
+    if (t == 0) {
+        int64_t run = 0;
+        for (int i = 0; i < (int)blockDim.x; ++i) {
+            const int64_t v = part[i];
+            part[i] = run;
+            run += v;
+        }
+        offsets[k] = run;
+    }
+    __syncthreads();
+    int64_t run = part[t];
+    for (int j = lo; j < hi; ++j) {
+        offsets[j] = run;
+        run += counts[j];
+        if (counts64) {
+            if (accumulate)
+                counts64[j] += counts[j];
+            else
+                counts64[j] = counts[j];
+        }
+    }
+}
+
+cudaError_t launch_scan_offsets(const int32_t *counts32, int k, int64_t *offsets,
+                                int64_t *counts64_out, int accumulate_counts, cudaStream_t st) {
+    scan_offsets_kernel<<<1, 1024, 0, st>>>(counts32, k, offsets, counts64_out,
+                                            accumulate_counts);
+    return launched();
+}
+
+// ------------------------------------------------------------------ scatter
+__global__ void scatter_kernel(const int32_t *__restrict__ assign, int64_t n, int k,
+                               const int64_t *__restrict__ offsets, int32_t *__restrict__ cursor,
+                               int32_t *__restrict__ perm) {
+    for (int64_t t = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; t < n;
+         t += (int64_t)gridDim.x * blockDim.x) {
+        const int a = assign[t];
+        if (a < 0 || a >= k) continue;  // skipped consistently with the histogram
+        const int pos = atomicAdd(&cursor[a], 1);
+        perm[offsets[a] + pos] = (int32_t)t;
+    }
+}
+
+cudaError_t launch_scatter(const int32_t *assign, int64_t n, int k, const int64_t *offsets,
+                           int32_t *cursor, int32_t *perm, cudaStream_t st) {
+    if (n == 0) return cudaSuccess;
+    int64_t blocks = (n + 255) / 256;
+    if (blocks > 152 * 8) blocks = 152 * 8;
+    scatter_kernel<<<(unsigned)blocks, 256, 0, st>>>(assign, n, k, offsets, cursor, perm);
+    return launched();
+}
+
+// ------------------------------------------------------ segmented sums: float
+// One CTA per cluster; thread t owns dimensions t, t + 256, ... (up to 16).
+// Members are read four at a time for memory-level parallelism.
+constexpr int SEG_THREADS = 256;
+constexpr int SEG_MAXV = 16;  // d <= 4096
+
+template <bool BF16>
+__global__ void __launch_bounds__(SEG_THREADS) segsum_float_kernel(
+    const void *__restrict__ Xv, int d, const int32_t *__restrict__ perm,
+    const int64_t *__restrict__ offsets, float *__restrict__ C, double *__restrict__ partial) {
+    const int j = blockIdx.x;
+    const int64_t lo = offsets[j], hi = offsets[j + 1];
+    const int64_t cnt = hi - lo;
+    if (cnt == 0) return;  // empty cluster keeps its centroid / adds nothing
+    float acc[SEG_MAXV];
+#pragma unroll
+    for (int v = 0; v < SEG_MAXV; ++v) acc[v] = 0.0f;
+    for (int64_t q = lo; q < hi; ++q) {
+        const int64_t p = perm[q];
+        if (BF16) {
+            const uint16_t *x = reinterpret_cast<const uint16_t *>(Xv) + p * d;
+#pragma unroll
+            for (int v = 0; v < SEG_MAXV; ++v) {
+                const int i = threadIdx.x + v * SEG_THREADS;
+                if (i < d) acc[v] += __uint_as_float(((uint32_t)__ldg(x + i)) << 16);
+            }
+        } else {
+            const float *x = reinterpret_cast<const float *>(Xv) + p * d;
+#pragma unroll
+            for (int v = 0; v < SEG_MAXV; ++v) {
+                const int i = threadIdx.x + v * SEG_THREADS;
+                if (i < d) acc[v] += __ldg(x + i);
+            }
+        }
+    }
+#pragma unroll
+    for (int v = 0; v < SEG_MAXV; ++v) {
+        const int i = threadIdx.x + v * SEG_THREADS;
+        if (i < d) {
+            if (partial)
+                partial[(int64_t)j * d + i] += (double)acc[v];
+            else
+                C[(int64_t)j * d + i] = __fdiv_rn(acc[v], (float)cnt);
+        }
+    }
+}
+
+cudaError_t launch_segsum_float(const void *X, int x_is_bf16, int d, const int32_t *perm,
+                                const int64_t *offsets, int k, float *C_inout, double *partial,
+                                cudaStream_t st) {
+    if (x_is_bf16)
+        segsum_float_kernel<true><<<k, SEG_THREADS, 0, st>>>(X, d, perm, offsets, C_inout, partial);
+    else
+        segsum_float_kernel<false><<<k, SEG_THREADS, 0, st>>>(X, d, perm, offsets, C_inout,
+                                                              partial);
+    return launched();
+}
+
+// ------------------------------------------------------- segmented sums: SQ8
+__device__ __forceinline__ uint8_t round_half_even_div(int64_t S, int64_t m) {
+    int64_t q = S / m;
+    const int64_t r = S - q * m;
+    if (2 * r > m || (2 * r == m && (q & 1))) q += 1;
+    return (uint8_t)q;
+}
+
+__global__ void __launch_bounds__(SEG_THREADS) segsum_sq8_kernel(
+    const uint8_t *__restrict__ X, int d, const int32_t *__restrict__ perm,
+    const int64_t *__restrict__ offsets, uint8_t *__restrict__ C, int64_t *__restrict__ partial) {
+    const int j = blockIdx.x;
+    const int64_t lo = offsets[j], hi = offsets[j + 1];
+    const int64_t cnt = hi - lo;
+    if (cnt == 0) return;
+    int64_t acc[SEG_MAXV];
+#pragma unroll
+    for (int v = 0; v < SEG_MAXV; ++v) acc[v] = 0;
+    for (int64_t q = lo; q < hi; ++q) {
+        const uint8_t *x = X + (int64_t)perm[q] * d;
+#pragma unroll
+        for (int v = 0; v < SEG_MAXV; ++v) {
+            const int i = threadIdx.x + v * SEG_THREADS;
+            if (i < d) acc[v] += __ldg(x + i);
+        }
+    }
+#pragma unroll
+    for (int v = 0; v < SEG_MAXV; ++v) {
+        const int i = threadIdx.x + v * SEG_THREADS;
+        if (i < d) {
+            if (partial)
+                partial[(int64_t)j * d + i] += acc[v];
+            else
+                C[(int64_t)j * d + i] = round_half_even_div(acc[v], cnt);
+        }
+    }
+}
+
+cudaError_t launch_segsum_sq8(const uint8_t *X, int d, const int32_t *perm,
+                              const int64_t *offsets, int k, uint8_t *C_inout, int64_t *partial,
+                              cudaStream_t st) {
+    segsum_sq8_kernel<<<k, SEG_THREADS, 0, st>>>(X, d, perm, offsets, C_inout, partial);
+    return launched();
+}
+
+// ------------------------------------------------------ segmented sums: RBQ1
+// Fused decode-average with exact fixed-point sums: Fq = rint(F 2^e),
+// T_i = sum Fq xbar_i, U = sum Fq;
+// c_i = m_i + (((2 T_i - U) 2^-e) / count) / sqrt(d) in fp64 -> fp32.
+__device__ __forceinline__ float rbq1_finish(int64_t T, int64_t U, int64_t cnt, float m,
+                                             double pow2m, double isd) {
+    double v = __ll2double_rn(2 * T - U);
+    v = __dmul_rn(v, pow2m);
+    v = __ddiv_rn(v, (double)cnt);
+    v = __dmul_rn(v, isd);
+    return __double2float_rn(__dadd_rn((double)m, v));
+}
+
+__global__ void __launch_bounds__(SEG_THREADS) segsum_rbq1_kernel(
+    const uint32_t *__restrict__ codes, const float *__restrict__ F, int d,
+    const float *__restrict__ m, int e, const int32_t *__restrict__ perm,
+    const int64_t *__restrict__ offsets, float *__restrict__ C, int64_t *__restrict__ partial) {
+    const int j = blockIdx.x;
+    const int64_t lo = offsets[j], hi = offsets[j + 1];
+    const int64_t cnt = hi - lo;
+    if (cnt == 0) return;
+    const int W = (d + 31) >> 5;
+    const double pow2 = ldexp(1.0, e);
+    int64_t acc[SEG_MAXV];
+#pragma unroll
+    for (int v = 0; v < SEG_MAXV; ++v) acc[v] = 0;
+    int64_t U = 0;
+    for (int64_t q = lo; q < hi; ++q) {
+        const int64_t p = perm[q];
+        const int64_t fq = __double2ll_rn(__dmul_rn((double)__ldg(F + p), pow2));
+        U += fq;
+        const uint32_t *cw = codes + p * W;
+#pragma unroll
+        for (int v = 0; v < SEG_MAXV; ++v) {
+            const int i = threadIdx.x + v * SEG_THREADS;
+            if (i < d) {
+                const uint32_t word = __ldg(cw + (i >> 5));
+                if ((word >> (i & 31)) & 1u) acc[v] += fq;
+            }
+        }
+    }
+    const double pow2m = ldexp(1.0, -e);
+    const double isd = __ddiv_rn(1.0, __dsqrt_rn((double)d));
+#pragma unroll
+    for (int v = 0; v < SEG_MAXV; ++v) {
+        const int i = threadIdx.x + v * SEG_THREADS;
+        if (i < d) {
+            if (partial)
+                partial[(int64_t)j * (d + 1) + i] += acc[v];
+            else
+                C[(int64_t)j * d + i] = rbq1_finish(acc[v], U, cnt, m[i], pow2m, isd);
+        }
+    }
+    if (partial && threadIdx.x == 0) partial[(int64_t)j * (d + 1) + d] += U;
+}
+
+cudaError_t launch_segsum_rbq1(const uint32_t *codes, const float *F, int d, const float *m,
+                               int e, const int32_t *perm, const int64_t *offsets, int k,
+                               float *C_inout, int64_t *partial, cudaStream_t st) {
+    segsum_rbq1_kernel<<<k, SEG_THREADS, 0, st>>>(codes, F, d, m, e, perm, offsets, C_inout,
+                                                  partial);
+    return launched();
+}
+
+// --------------------------------------------------------------- finalizers
+__global__ void finalize_float_kernel(const double *__restrict__ partial,
+                                      const int64_t *__restrict__ counts, int k, int d,
+                                      float *__restrict__ C) {
+    const int64_t t = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
+    if (t >= (int64_t)k * d) return;
+    const int j = (int)(t / d);
+    const int64_t c = counts[j];
+    if (c > 0) C[t] = __double2float_rn(__ddiv_rn(partial[t], (double)c));
+}
+
+cudaError_t launch_finalize_float(const double *partial, const int64_t *counts, int k, int d,
+                                  float *C_inout, cudaStream_t st) {
+    const int64_t tot = (int64_t)k * d;
+    finalize_float_kernel<<<(unsigned)((tot + 255) / 256), 256, 0, st>>>(partial, counts, k, d,
+                                                                         C_inout);
+    return launched();
+}
+
+__global__ void finalize_sq8_kernel(const int64_t *__restrict__ partial,
+                                    const int64_t *__restrict__ counts, int k, int d,
+                                    uint8_t *__restrict__ C) {
+    const int64_t t = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
+    if (t >= (int64_t)k * d) return;
+    const int j = (int)(t / d);
+    const int64_t c = counts[j];
+    if (c > 0) C[t] = round_half_even_div(partial[t], c);
+}
+
+cudaError_t launch_finalize_sq8(const int64_t *partial, const int64_t *counts, int k, int d,
+                                uint8_t *C_inout, cudaStream_t st) {
+    const int64_t tot = (int64_t)k * d;
+    finalize_sq8_kernel<<<(unsigned)((tot + 255) / 256), 256, 0, st>>>(partial, counts, k, d,
+                                                                       C_inout);
+    return launched();
+}
+
+__global__ void finalize_rbq1_kernel(const int64_t *__restrict__ partial,
+                                     const int64_t *__restrict__ counts, int k, int d,
+                                     const float *__restrict__ m, int e, float *__restrict__ C) {
+    const int64_t t = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
+    if (t >= (int64_t)k * d) return;
+    const int j = (int)(t / d), i = (int)(t - (int64_t)j * d);
+    const int64_t c = counts[j];
+    if (c <= 0) return;
+    const double pow2m = ldexp(1.0, -e);
+    const double isd = __ddiv_rn(1.0, __dsqrt_rn((double)d));
+    C[t] = rbq1_finish(partial[(int64_t)j * (d + 1) + i], partial[(int64_t)j * (d + 1) + d], c,
+                       m[i], pow2m, isd);
+}
+
+cudaError_t launch_finalize_rbq1(const int64_t *partial, const int64_t *counts, int k, int d,
+                                 const float *m, int e, float *C_inout, cudaStream_t st) {
+    const int64_t tot = (int64_t)k * d;
+    finalize_rbq1_kernel<<<(unsigned)((tot + 255) / 256), 256, 0, st>>>(partial, counts, k, d, m,
+                                                                        e, C_inout);
+    return launched();
+}
+
+__global__ void merge_kernel(void *__restrict__ dst, const void *__restrict__ src, int64_t count,
+                             int elem_type) {
+    for (int64_t t = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; t < count;
+         t += (int64_t)gridDim.x * blockDim.x) {
+        if (elem_type == 0)
+            reinterpret_cast<double *>(dst)[t] += reinterpret_cast<const double *>(src)[t];
+        else
+            reinterpret_cast<int64_t *>(dst)[t] += reinterpret_cast<const int64_t *>(src)[t];
+    }
+}
+
+cudaError_t launch_merge(void *dst, const void *src, int64_t count, int elem_type,
+                         cudaStream_t st) {
+    if (count == 0) return cudaSuccess;
+    int64_t blocks = (count + 255) / 256;
+    if (blocks > 152 * 8) blocks = 152 * 8;
+    merge_kernel<<<(unsigned)blocks, 256, 0, st>>>(dst, src, count, elem_type);
+    return launched();
+}
+
+}  // namespace skm

@@ -1,0 +1,553 @@
+// extern "C" entry points of libskm (declared in include/skm.h): argument
+// validation on the host, workspace carving, and the launch sequences of the
+// Lloyd k-means hot path (Section 2.3) for each representation.
+#include <stdarg.h>
+#include <stdio.h>
+
+#include <algorithm>
+#include <atomic>
+#include <cmath>
+#include <vector>
+
+#include "skm_internal.cuh"
+#include "skm_tc.cuh"
+
+namespace skm {
+
+static thread_local char g_err[512] = "";
+static std::atomic<unsigned long long> g_launches{0};
+
+cudaError_t launched(int count) {
+    g_launches.fetch_add((unsigned long long)count, std::memory_order_relaxed);
+    return cudaGetLastError();
+}
+
+int set_error(int code, const char *fmt, ...) {
+    va_list ap;
+    va_start(ap, fmt);
+    vsnprintf(g_err, sizeof(g_err), fmt, ap);
+    va_end(ap);
+    return code;
+}
+
+static inline cudaStream_t S(void *s) { return static_cast<cudaStream_t>(s); }
+
+constexpr int MAX_D = 4096;
+constexpr int MAX_K = 65536;
+constexpr int64_t MAX_N = (int64_t(1) << 31) - 1;
+constexpr int64_t MAX_N_RBQ1 = int64_t(1) << 24;
+constexpr int RED_BLOCKS = 304;  // 2 x 152 SMs for column / objective reductions
+
+static int check_data(const skm_data *x, bool need_codes = true) {
+    if (!x) return set_error(SKM_ERR_INVALID_ARG, "skm_data is NULL");
+    if (x->repr < SKM_REPR_F32 || x->repr > SKM_REPR_BF16)
+        return set_error(SKM_ERR_INVALID_ARG, "unknown repr %d", x->repr);
+    if (x->d < 1 || x->d > MAX_D)
+        return set_error(x->d < 1 ? SKM_ERR_INVALID_ARG : SKM_ERR_UNSUPPORTED,
+                         "d = %d outside [1, %d]", x->d, MAX_D);
+    if (x->n < 1 || x->n > MAX_N)
+        return set_error(x->n < 1 ? SKM_ERR_INVALID_ARG : SKM_ERR_UNSUPPORTED,
+                         "n = %lld outside [1, 2^31)", (long long)x->n);
+    if (need_codes && !x->x) return set_error(SKM_ERR_INVALID_ARG, "x->x is NULL");
+    if (x->repr == SKM_REPR_RBQ1) {
+        if (x->n > MAX_N_RBQ1)
+            return set_error(SKM_ERR_UNSUPPORTED, "RBQ1 supports n <= 2^24 (got %lld)",
+                             (long long)x->n);
+        if (!x->nx2 || !x->F || !x->popx || !x->m)
+            return set_error(SKM_ERR_INVALID_ARG, "RBQ1 needs nx2, F, popx and m");
+    }
+    return SKM_OK;
+}
+
+static int check_k(const skm_data *x, int k) {
+    if (k < 1 || k > MAX_K)
+        return set_error(k < 1 ? SKM_ERR_INVALID_ARG : SKM_ERR_UNSUPPORTED,
+                         "k = %d outside [1, %d]", k, MAX_K);
+    if ((int64_t)k > x->n)
+        return set_error(SKM_ERR_INVALID_ARG, "k = %d exceeds n = %lld", k, (long long)x->n);
+    return SKM_OK;
+}
+
+// ------------------------------------------------------------ workspace plans
+struct AssignBufs {
+    int32_t *nx = nullptr, *nc = nullptr;  // SQ8
+    uint4 *planes = nullptr;                // RBQ1
+    Rbq1CInfo *info = nullptr;
+    TcAssignBufs tc;                        // F32 / BF16 / SQ8 tensor-core screen
+};
+
+static void plan_assign(const skm_data *x, int k, Carver &cv, AssignBufs &b) {
+    const int64_t n = x->n;
+    const int d = x->d;
+    switch (x->repr) {
+    case SKM_REPR_SQ8:
+        b.nx = cv.take<int32_t>(n);
+        b.nc = cv.take<int32_t>(k);
+        break;
+    case SKM_REPR_RBQ1:
+        b.planes = cv.take<uint4>((size_t)k * words_of(d));
+        b.info = cv.take<Rbq1CInfo>(k);
+        break;
+    default:
+        break;
+    }
+    tc_plan(x->repr, n, d, k, cv, b.tc);
+}
+
+struct UpdateBufs {
+    int32_t *counts32 = nullptr, *cursor = nullptr, *perm = nullptr;
+    int64_t *offsets = nullptr;
+};
+
+static void plan_update(const skm_data *x, int k, Carver &cv, UpdateBufs &b) {
+    b.counts32 = cv.take<int32_t>(k);
+    b.cursor = cv.take<int32_t>(k);
+    b.offsets = cv.take<int64_t>((size_t)k + 1);
+    b.perm = cv.take<int32_t>(x->n);
+}
+
+struct FitBufs {
+    AssignBufs a;
+    UpdateBufs u;
+    float *dist = nullptr;
+    double *partials = nullptr, *sum = nullptr;
+    unsigned int *maxbits = nullptr;
+    int *e_dev = nullptr;
+    int *status = nullptr;
+    int64_t *counts = nullptr;
+};
+
+static void plan_fit(const skm_data *x, int k, Carver &cv, FitBufs &b) {
+    plan_assign(x, k, cv, b.a);
+    plan_update(x, k, cv, b.u);
+    b.dist = cv.take<float>(x->n);
+    b.partials = cv.take<double>(RED_BLOCKS);
+    b.sum = cv.take<double>(1);
+    b.maxbits = cv.take<unsigned int>(1);
+    b.e_dev = cv.take<int>(1);
+    b.status = cv.take<int>(1);
+    b.counts = cv.take<int64_t>(k);
+}
+
+static int need_ws(const Carver &cv, size_t ws_bytes, void *ws) {
+    if (cv.off > ws_bytes)
+        return set_error(SKM_ERR_NO_MEMORY, "workspace too small: need %zu bytes, got %zu", cv.off,
+                         ws_bytes);
+    if (cv.off > 0 && !ws) return set_error(SKM_ERR_INVALID_ARG, "workspace is NULL");
+    if (((uintptr_t)ws & 255) != 0)
+        return set_error(SKM_ERR_INVALID_ARG, "workspace must be 256-byte aligned");
+    return SKM_OK;
+}
+
+// ------------------------------------------------------------ core steps
+static int do_assign(const skm_data *x, const void *C, int k, const int32_t *prev,
+                     int32_t *assign, float *dist, AssignBufs &b, cudaStream_t st) {
+    const int64_t n = x->n;
+    const int d = x->d;
+    switch (x->repr) {
+    case SKM_REPR_F32:
+        SKM_TRY(tc_assign_float(x, static_cast<const float *>(C), k, assign, dist, b.tc, st));
+        break;
+    case SKM_REPR_BF16:
+        SKM_TRY(tc_assign_float(x, static_cast<const float *>(C), k, assign, dist, b.tc, st));
+        (void)prev;
+        break;
+    case SKM_REPR_SQ8: {
+        const uint8_t *X = static_cast<const uint8_t *>(x->x);
+        const uint8_t *Cc = static_cast<const uint8_t *>(C);
+        SKM_CUDA_TRY(launch_row_sqnorm_u8(X, n, d, b.nx, st));
+        SKM_CUDA_TRY(launch_row_sqnorm_u8(Cc, k, d, b.nc, st));
+        SKM_TRY(tc_assign_sq8(x, Cc, k, b.nx, b.nc, assign, dist, b.tc, st));
+        break;
+    }
+    case SKM_REPR_RBQ1:
+        SKM_CUDA_TRY(
+            launch_rbq1_cprep(static_cast<const float *>(C), k, d, x->m, b.planes, b.info, st));
+        SKM_CUDA_TRY(launch_assign_rbq1(static_cast<const uint32_t *>(x->x), x->nx2, x->F, x->popx,
+                                        n, d, b.planes, b.info, k, assign, dist, st));
+        break;
+    }
+    return SKM_OK;
+}
+
+static int do_update(const skm_data *x, const int32_t *assign, int k, void *C, int64_t *counts,
+                     void *partial, int e, UpdateBufs &b, cudaStream_t st) {
+    const int64_t n = x->n;
+    const int d = x->d;
+    SKM_CUDA_TRY(launch_histogram(assign, n, k, b.counts32, st));
+    SKM_CUDA_TRY(launch_scan_offsets(b.counts32, k, b.offsets, counts, partial ? 1 : 0, st));
+    SKM_CUDA_TRY(cudaMemsetAsync(b.cursor, 0, sizeof(int32_t) * (size_t)k, st));
+    SKM_CUDA_TRY(launch_scatter(assign, n, k, b.offsets, b.cursor, b.perm, st));
+    switch (x->repr) {
+    case SKM_REPR_F32:
+    case SKM_REPR_BF16:
+        SKM_CUDA_TRY(launch_segsum_float(x->x, x->repr == SKM_REPR_BF16, d, b.perm, b.offsets, k,
+                                         static_cast<float *>(C), static_cast<double *>(partial),
+                                         st));
+        break;
+    case SKM_REPR_SQ8:
+        SKM_CUDA_TRY(launch_segsum_sq8(static_cast<const uint8_t *>(x->x), d, b.perm, b.offsets, k,
+                                       static_cast<uint8_t *>(C), static_cast<int64_t *>(partial),
+                                       st));
+        break;
+    case SKM_REPR_RBQ1:
+        SKM_CUDA_TRY(launch_segsum_rbq1(static_cast<const uint32_t *>(x->x), x->F, d, x->m, e,
+                                        b.perm, b.offsets, k, static_cast<float *>(C),
+                                        static_cast<int64_t *>(partial), st));
+        break;
+    }
+    return SKM_OK;
+}
+
+static size_t centroid_bytes(const skm_data *x, int k) {
+    return (size_t)k * x->d * (x->repr == SKM_REPR_SQ8 ? 1 : 4);
+}
+
+}  // namespace skm
+
+using namespace skm;
+
+extern "C" {
+
+const char *skm_last_error(void) { return g_err; }
+
+int skm_version(void) { return 100; }
+
+uint64_t skm_kernel_launches(void) { return (uint64_t)g_launches.load(std::memory_order_relaxed); }
+
+size_t skm_workspace_size(int op, const skm_data *x, int k) {
+    Carver cv(nullptr, 0);
+    switch (op) {
+    case 0: {
+        if (check_data(x, false) || check_k(x, k)) return 0;
+        AssignBufs b;
+        plan_assign(x, k, cv, b);
+        break;
+    }
+    case 1: {
+        if (check_data(x, false) || check_k(x, k)) return 0;
+        UpdateBufs b;
+        plan_update(x, k, cv, b);
+        break;
+    }
+    case 2: {
+        if (check_data(x, false) || check_k(x, k)) return 0;
+        FitBufs b;
+        plan_fit(x, k, cv, b);
+        break;
+    }
+    case 3: {  // quantize: column reductions
+        if (!x || x->d < 1 || x->d > MAX_D) {
+            set_error(SKM_ERR_INVALID_ARG, "bad skm_data for op 3");
+            return 0;
+        }
+        cv.take<double>((size_t)RED_BLOCKS * x->d);
+        cv.take<float>((size_t)RED_BLOCKS * x->d);
+        cv.take<float>((size_t)RED_BLOCKS * x->d);
+        cv.take<unsigned int>(1);
+        cv.take<int>(1);
+        break;
+    }
+    case 4: {  // pca
+        if (!x || x->d < 1 || x->d > MAX_D) {
+            set_error(SKM_ERR_INVALID_ARG, "bad skm_data for op 4");
+            return 0;
+        }
+        const int d = x->d;
+        const int splits = 32;
+        cv.take<double>((size_t)RED_BLOCKS * d);
+        cv.take<double>((size_t)splits * d * d);
+        cv.take<double>((size_t)d * d);
+        break;
+    }
+    default:
+        set_error(SKM_ERR_INVALID_ARG, "unknown op %d", op);
+        return 0;
+    }
+    return cv.off < 256 ? 256 : cv.off;
+}
+
+int skm_project(const float *X, int64_t n, int d, const float *mean, const float *P, int d_out,
+                int out_dtype, void *Y, void *stream) {
+    if (!X || !P || !Y) return set_error(SKM_ERR_INVALID_ARG, "NULL pointer");
+    if (n < 1 || d < 1 || d > MAX_D || d_out < 1 || d_out > d)
+        return set_error(SKM_ERR_INVALID_ARG, "bad shape n=%lld d=%d d_out=%d", (long long)n, d,
+                         d_out);
+    if (out_dtype != SKM_DTYPE_F32 && out_dtype != SKM_DTYPE_BF16)
+        return set_error(SKM_ERR_INVALID_ARG, "bad out_dtype %d", out_dtype);
+    SKM_CUDA_TRY(launch_project(X, n, d, mean, P, d_out, out_dtype == SKM_DTYPE_BF16, Y,
+                                S(stream)));
+    return SKM_OK;
+}
+
+int skm_make_rotation(uint64_t seed, int d, float *P_host) {
+    if (!P_host || d < 1 || d > MAX_D) return set_error(SKM_ERR_INVALID_ARG, "bad arguments");
+    std::vector<double> A((size_t)d * d);
+    philox_gaussians(seed, (int64_t)d * d, A.data());
+    householder_qr_q(d, A.data());
+    for (size_t i = 0; i < A.size(); ++i) P_host[i] = (float)A[i];
+    return SKM_OK;
+}
+
+int skm_pca_fit(const float *X, int64_t n, int d, int d_out, float *mean, float *P,
+                float *eigvals, void *ws, size_t ws_bytes, void *stream) {
+    if (!X || !mean || !P) return set_error(SKM_ERR_INVALID_ARG, "NULL pointer");
+    if (n < 2 || d < 1 || d > MAX_D || d_out < 1 || d_out > d)
+        return set_error(SKM_ERR_INVALID_ARG, "bad shape");
+    cudaStream_t st = S(stream);
+    const int splits = 32;
+    Carver cv(ws, ws_bytes);
+    double *psum = cv.take<double>((size_t)RED_BLOCKS * d);
+    double *partial = cv.take<double>((size_t)splits * d * d);
+    double *cov = cv.take<double>((size_t)d * d);
+    SKM_TRY(need_ws(cv, ws_bytes, ws));
+    const int nblk = (int)std::min<int64_t>(RED_BLOCKS, n);
+    SKM_CUDA_TRY(launch_colsum_partial(X, n, d, psum, nblk, st));
+    SKM_CUDA_TRY(launch_colmean_finish(psum, nblk, d, n, mean, nullptr, st));
+    SKM_CUDA_TRY(launch_cov_partial(X, n, d, mean, partial, splits, st));
+    SKM_CUDA_TRY(launch_cov_reduce(partial, splits, d, cov, st));
+    std::vector<double> A((size_t)d * d), w(d);
+    SKM_CUDA_TRY(cudaMemcpyAsync(A.data(), cov, sizeof(double) * A.size(), cudaMemcpyDeviceToHost,
+                                 st));
+    SKM_CUDA_TRY(cudaStreamSynchronize(st));
+    for (auto &v : A) v /= (double)n;
+    if (symmetric_eigen(d, A.data(), w.data()) != 0)
+        return set_error(SKM_ERR_UNSUPPORTED, "eigen-decomposition did not converge");
+    std::vector<int> order(d);
+    for (int i = 0; i < d; ++i) order[i] = i;
+    std::stable_sort(order.begin(), order.end(), [&](int a, int b) { return w[a] > w[b]; });
+    std::vector<float> Ph((size_t)d * d_out), wh(d_out);
+    for (int j = 0; j < d_out; ++j) {
+        const int c = order[j];
+        int piv = 0;
+        for (int i = 1; i < d; ++i)
+            if (fabs(A[(size_t)i * d + c]) > fabs(A[(size_t)piv * d + c])) piv = i;
+        const double sg = A[(size_t)piv * d + c] < 0 ? -1.0 : 1.0;
+        for (int i = 0; i < d; ++i) Ph[(size_t)i * d_out + j] = (float)(sg * A[(size_t)i * d + c]);
+        wh[j] = (float)w[c];
+    }
+    SKM_CUDA_TRY(cudaMemcpyAsync(P, Ph.data(), sizeof(float) * Ph.size(), cudaMemcpyHostToDevice,
+                                 st));
+    if (eigvals)
+        SKM_CUDA_TRY(cudaMemcpyAsync(eigvals, wh.data(), sizeof(float) * wh.size(),
+                                     cudaMemcpyHostToDevice, st));
+    SKM_CUDA_TRY(cudaStreamSynchronize(st));
+    return SKM_OK;
+}
+
+int skm_quantize(int repr, const float *X, int64_t n, int d, skm_quant_params *qp, void *codes,
+                 void *ws, size_t ws_bytes, void *stream) {
+    if (!X || !qp || !codes) return set_error(SKM_ERR_INVALID_ARG, "NULL pointer");
+    if (n < 1 || n > MAX_N || d < 1 || d > MAX_D)
+        return set_error(SKM_ERR_INVALID_ARG, "bad shape n=%lld d=%d", (long long)n, d);
+    cudaStream_t st = S(stream);
+    Carver cv(ws, ws_bytes);
+    double *psum = cv.take<double>((size_t)RED_BLOCKS * d);
+    float *pmin = cv.take<float>((size_t)RED_BLOCKS * d);
+    float *pmax = cv.take<float>((size_t)RED_BLOCKS * d);
+    const int nblk = (int)std::min<int64_t>(RED_BLOCKS, n);
+    if (repr == SKM_REPR_SQ8) {
+        if (!qp->b || !qp->s) return set_error(SKM_ERR_INVALID_ARG, "SQ8 needs b and s");
+        if (qp->fit) {
+            SKM_TRY(need_ws(cv, ws_bytes, ws));
+            SKM_CUDA_TRY(launch_colminmax_partial(X, n, d, pmin, pmax, nblk, st));
+            SKM_CUDA_TRY(launch_sq8_params(pmin, pmax, nblk, d, qp->b, qp->s, st));
+        }
+        SKM_CUDA_TRY(launch_sq8_encode(X, n, d, qp->b, qp->s, static_cast<uint8_t *>(codes), st));
+        return SKM_OK;
+    }
+    if (repr == SKM_REPR_RBQ1) {
+        if (n > MAX_N_RBQ1) return set_error(SKM_ERR_UNSUPPORTED, "RBQ1 supports n <= 2^24");
+        if (!qp->m || !qp->nx2 || !qp->F || !qp->popx)
+            return set_error(SKM_ERR_INVALID_ARG, "RBQ1 needs m, nx2, F and popx");
+        if (qp->fit) {
+            SKM_TRY(need_ws(cv, ws_bytes, ws));
+            SKM_CUDA_TRY(launch_colsum_partial(X, n, d, psum, nblk, st));
+            SKM_CUDA_TRY(launch_colmean_finish(psum, nblk, d, n, qp->m, nullptr, st));
+        }
+        SKM_CUDA_TRY(launch_rbq1_encode(X, n, d, qp->m, static_cast<uint32_t *>(codes), qp->nx2,
+                                        qp->F, qp->popx, st));
+        return SKM_OK;
+    }
+    return set_error(SKM_ERR_INVALID_ARG, "skm_quantize: repr must be SQ8 or RBQ1");
+}
+
+int skm_rbq1_exponent(const float *F, int64_t n, int *e_host, void *ws, size_t ws_bytes,
+                      void *stream) {
+    if (!F || !e_host || n < 1) return set_error(SKM_ERR_INVALID_ARG, "bad arguments");
+    cudaStream_t st = S(stream);
+    Carver cv(ws, ws_bytes);
+    unsigned int *mb = cv.take<unsigned int>(1);
+    int *ed = cv.take<int>(1);
+    SKM_TRY(need_ws(cv, ws_bytes, ws));
+    SKM_CUDA_TRY(launch_rbq1_exponent(F, n, mb, ed, st));
+    SKM_CUDA_TRY(cudaMemcpyAsync(e_host, ed, sizeof(int), cudaMemcpyDeviceToHost, st));
+    SKM_CUDA_TRY(cudaStreamSynchronize(st));
+    return SKM_OK;
+}
+
+int skm_assign(const skm_data *x, const void *C, int k, const int32_t *prev_assign,
+               int32_t *assign, float *dist, void *ws, size_t ws_bytes, void *stream) {
+    SKM_TRY(check_data(x));
+    SKM_TRY(check_k(x, k));
+    if (!C || !assign) return set_error(SKM_ERR_INVALID_ARG, "C and assign are required");
+    Carver cv(ws, ws_bytes);
+    AssignBufs b;
+    plan_assign(x, k, cv, b);
+    SKM_TRY(need_ws(cv, ws_bytes, ws));
+    return do_assign(x, C, k, prev_assign, assign, dist, b, S(stream));
+}
+
+int skm_update(const skm_data *x, const int32_t *assign, int k, void *C_inout, int64_t *counts,
+               void *partial, void *ws, size_t ws_bytes, void *stream) {
+    SKM_TRY(check_data(x));
+    SKM_TRY(check_k(x, k));
+    if (!assign || !counts || (!C_inout && !partial))
+        return set_error(SKM_ERR_INVALID_ARG, "assign, counts and C_inout/partial are required");
+    Carver cv(ws, ws_bytes);
+    UpdateBufs b;
+    plan_update(x, k, cv, b);
+    SKM_TRY(need_ws(cv, ws_bytes, ws));
+    return do_update(x, assign, k, C_inout, counts, partial, x->rbq1_exp, b, S(stream));
+}
+
+int skm_merge_partials(void *dst, const void *src, int64_t count, int elem_type, void *stream) {
+    if (!dst || !src || count < 0 || (elem_type != 0 && elem_type != 1))
+        return set_error(SKM_ERR_INVALID_ARG, "bad arguments");
+    SKM_CUDA_TRY(launch_merge(dst, src, count, elem_type, S(stream)));
+    return SKM_OK;
+}
+
+int skm_update_finalize(const skm_data *x, const void *partial, const int64_t *counts, int k,
+                        void *C_inout, void *stream) {
+    SKM_TRY(check_data(x, false));
+    if (!partial || !counts || !C_inout || k < 1)
+        return set_error(SKM_ERR_INVALID_ARG, "bad arguments");
+    cudaStream_t st = S(stream);
+    switch (x->repr) {
+    case SKM_REPR_F32:
+    case SKM_REPR_BF16:
+        SKM_CUDA_TRY(launch_finalize_float(static_cast<const double *>(partial), counts, k, x->d,
+                                           static_cast<float *>(C_inout), st));
+        break;
+    case SKM_REPR_SQ8:
+        SKM_CUDA_TRY(launch_finalize_sq8(static_cast<const int64_t *>(partial), counts, k, x->d,
+                                         static_cast<uint8_t *>(C_inout), st));
+        break;
+    case SKM_REPR_RBQ1:
+        if (!x->m) return set_error(SKM_ERR_INVALID_ARG, "RBQ1 finalize needs m");
+        SKM_CUDA_TRY(launch_finalize_rbq1(static_cast<const int64_t *>(partial), counts, k, x->d,
+                                          x->m, x->rbq1_exp, static_cast<float *>(C_inout), st));
+        break;
+    }
+    return SKM_OK;
+}
+
+int skm_fit(const skm_fit_config *cfg, const skm_data *x, const void *C_init,
+            const int64_t *init_idx, void *C_out, int32_t *assign_out, float *dist_out,
+            double *objective_host, skm_stats *stats_host, void *ws, size_t ws_bytes,
+            void *stream) {
+    if (!cfg) return set_error(SKM_ERR_INVALID_ARG, "cfg is NULL");
+    SKM_TRY(check_data(x));
+    const int k = cfg->k;
+    SKM_TRY(check_k(x, k));
+    if (cfg->iters < 0 || cfg->iters > 100000)
+        return set_error(SKM_ERR_INVALID_ARG, "iters = %d", cfg->iters);
+    if (!C_out || !assign_out) return set_error(SKM_ERR_INVALID_ARG, "C_out and assign_out required");
+    if (!C_init && !init_idx)
+        return set_error(SKM_ERR_INVALID_ARG, "one of C_init / init_idx is required");
+    cudaStream_t st = S(stream);
+    Carver cv(ws, ws_bytes);
+    FitBufs b;
+    plan_fit(x, k, cv, b);
+    SKM_TRY(need_ws(cv, ws_bytes, ws));
+    const int64_t n = x->n;
+    const int d = x->d;
+
+    skm_data xd = *x;
+    int e = 0;
+    if (x->repr == SKM_REPR_RBQ1) {
+        SKM_CUDA_TRY(launch_rbq1_exponent(x->F, n, b.maxbits, b.e_dev, st));
+        SKM_CUDA_TRY(cudaMemcpyAsync(&e, b.e_dev, sizeof(int), cudaMemcpyDeviceToHost, st));
+        SKM_CUDA_TRY(cudaStreamSynchronize(st));
+        xd.rbq1_exp = e;
+    }
+    // STEP 1: initial centroids
+    SKM_CUDA_TRY(cudaMemsetAsync(b.status, 0, sizeof(int), st));
+    if (C_init) {
+        SKM_CUDA_TRY(cudaMemcpyAsync(C_out, C_init, centroid_bytes(x, k), cudaMemcpyDeviceToDevice,
+                                     st));
+    } else if (x->repr == SKM_REPR_RBQ1) {
+        SKM_CUDA_TRY(launch_rbq1_decode_rows(static_cast<const uint32_t *>(x->x), x->F, n, d, x->m,
+                                             e, init_idx, k, static_cast<float *>(C_out), b.status,
+                                             st));
+    } else {
+        const int eb = x->repr == SKM_REPR_SQ8 ? 1 : (x->repr == SKM_REPR_BF16 ? 2 : 4);
+        if (x->repr == SKM_REPR_BF16)
+            return set_error(SKM_ERR_INVALID_ARG, "BF16 fit needs fp32 C_init");
+        SKM_CUDA_TRY(launch_gather_rows(x->x, n, eb, d, init_idx, k, C_out, b.status, st));
+    }
+    if (!C_init) {
+        int bad = 0;
+        SKM_CUDA_TRY(cudaMemcpyAsync(&bad, b.status, sizeof(int), cudaMemcpyDeviceToHost, st));
+        SKM_CUDA_TRY(cudaStreamSynchronize(st));
+        if (bad) return set_error(SKM_ERR_DEVICE_CHECK, "init_idx holds an index outside [0, n)");
+    }
+    float *dist = dist_out ? dist_out : b.dist;
+    const int nblk = (int)std::min<int64_t>(RED_BLOCKS, n);
+    int32_t *assign = assign_out;
+    for (int it = 0; it <= cfg->iters; ++it) {
+        const bool want_obj = objective_host != nullptr;
+        SKM_TRY(do_assign(&xd, C_out, k, nullptr, assign, (want_obj || it == cfg->iters) ? dist
+                                                                                          : nullptr,
+                          b.a, st));
+        if (want_obj) {
+            SKM_CUDA_TRY(launch_sum_float_to_double(dist, n, b.partials, nblk, st));
+            SKM_CUDA_TRY(launch_sum_double(b.partials, nblk, b.sum, st));
+            SKM_CUDA_TRY(cudaMemcpyAsync(&objective_host[it], b.sum, sizeof(double),
+                                         cudaMemcpyDeviceToHost, st));
+        }
+        if (it == cfg->iters) break;
+        SKM_TRY(do_update(&xd, assign, k, C_out, b.counts, nullptr, e, b.u, st));
+    }
+    SKM_CUDA_TRY(cudaStreamSynchronize(st));
+    if (stats_host) {
+        memset(stats_host, 0, sizeof(*stats_host));
+        tc_read_stats(b.a.tc, stats_host, st);
+        std::vector<int64_t> cnt(k);
+        if (cfg->iters > 0) {
+            SKM_CUDA_TRY(cudaMemcpy(cnt.data(), b.counts, sizeof(int64_t) * k,
+                                    cudaMemcpyDeviceToHost));
+            for (int j = 0; j < k; ++j) stats_host->empty_clusters += cnt[j] == 0;
+        }
+    }
+    return SKM_OK;
+}
+
+int skm_objective(const void *X, int x_is_bf16, int64_t n, int d, const float *C, int k,
+                  const int32_t *assign, double *out_host, void *ws, size_t ws_bytes,
+                  void *stream) {
+    if (!X || !C || !assign || !out_host) return set_error(SKM_ERR_INVALID_ARG, "NULL pointer");
+    if (n < 1 || d < 1 || d > MAX_D || k < 1) return set_error(SKM_ERR_INVALID_ARG, "bad shape");
+    cudaStream_t st = S(stream);
+    Carver cv(ws, ws_bytes);
+    double *partials = cv.take<double>(RED_BLOCKS);
+    double *sum = cv.take<double>(1);
+    SKM_TRY(need_ws(cv, ws_bytes, ws));
+    const int nblk = (int)std::min<int64_t>(RED_BLOCKS, n);
+    SKM_CUDA_TRY(launch_objective(X, x_is_bf16, n, d, C, assign, partials, nblk, st));
+    SKM_CUDA_TRY(launch_sum_double(partials, nblk, sum, st));
+    SKM_CUDA_TRY(cudaMemcpyAsync(out_host, sum, sizeof(double), cudaMemcpyDeviceToHost, st));
+    SKM_CUDA_TRY(cudaStreamSynchronize(st));
+    return SKM_OK;
+}
+
+int skm_sq8_decode(const uint8_t *codes, int64_t n, int d, const float *b, const float *s,
+                   float *Y, void *stream) {
+    if (!codes || !b || !s || !Y || n < 1 || d < 1 || d > MAX_D)
+        return set_error(SKM_ERR_INVALID_ARG, "bad arguments");
+    SKM_CUDA_TRY(launch_sq8_decode(codes, n, d, b, s, Y, S(stream)));
+    return SKM_OK;
+}
+
+}  // extern "C"

@@ -1,0 +1,152 @@
+// Internal declarations shared by the libskm translation units (not part of
+// the ABI).  Kernels are launched through the `launch_*` functions declared
+// here; every launcher returns cudaGetLastError() of its launch.
+#pragma once
+
+#include <cuda_runtime.h>
+#include <cuda_bf16.h>
+#include <stdint.h>
+#include <stddef.h>
+
+#include "../../include/skm.h"
+
+namespace skm {
+
+// ---- error reporting (thread-local message, see skm_abi.cu) --------------
+int set_error(int code, const char *fmt, ...);
+
+#define SKM_CUDA_TRY(expr)                                                         \
+    do {                                                                           \
+        cudaError_t e_ = (expr);                                                   \
+        if (e_ != cudaSuccess)                                                     \
+            return ::skm::set_error(SKM_ERR_CUDA, "%s failed: %s (%s:%d)", #expr,  \
+                                    cudaGetErrorString(e_), __FILE__, __LINE__);   \
+    } while (0)
+
+#define SKM_TRY(expr)                    \
+    do {                                 \
+        int s_ = (expr);                 \
+        if (s_ != SKM_OK) return s_;     \
+    } while (0)
+
+// Counts `count` kernel launches (host-side, process-wide) and returns
+// cudaGetLastError(); every launcher returns through it.
+cudaError_t launched(int count = 1);
+
+// ---- workspace carving ------------------------------------------------------
+// Sub-buffers are carved from the caller's workspace at 256-byte boundaries.
+// With base == nullptr the carver only measures (used by skm_workspace_size).
+struct Carver {
+    char *base;
+    size_t off = 0;
+    size_t cap;
+    Carver(void *b, size_t c) : base(static_cast<char *>(b)), cap(c) {}
+    template <typename T>
+    T *take(size_t count) {
+        off = (off + 255) & ~size_t(255);
+        T *p = base ? reinterpret_cast<T *>(base + off) : nullptr;
+        off += count * sizeof(T);
+        return p;
+    }
+    bool fits() const { return off <= cap; }
+};
+
+inline int words_of(int d) { return (d + 31) / 32; }
+inline int64_t cdiv(int64_t a, int64_t b) { return (a + b - 1) / b; }
+
+// Per-centroid terms of the RBQ1 estimator (Eq. final:rabitq), one record
+// per centroid: SQ4 bias b, scale s, sum of codes, ||c - m||^2.
+struct Rbq1CInfo {
+    float b;
+    float s;
+    int32_t sumy;
+    float ny2;
+};
+
+// ---- kernels (launchers) ------------------------------------------------
+// quantize / encode
+cudaError_t launch_colminmax_partial(const float *X, int64_t n, int d, float *pmin, float *pmax,
+                                     int nblk, cudaStream_t st);
+cudaError_t launch_sq8_params(const float *pmin, const float *pmax, int nblk, int d, float *b,
+                              float *s, cudaStream_t st);
+cudaError_t launch_sq8_encode(const float *X, int64_t n, int d, const float *b, const float *s,
+                              uint8_t *codes, cudaStream_t st);
+cudaError_t launch_sq8_decode(const uint8_t *codes, int64_t n, int d, const float *b,
+                              const float *s, float *Y, cudaStream_t st);
+cudaError_t launch_colsum_partial(const float *X, int64_t n, int d, double *psum, int nblk,
+                                  cudaStream_t st);
+cudaError_t launch_colmean_finish(const double *psum, int nblk, int d, int64_t n, float *m,
+                                  double *mean_d, cudaStream_t st);
+cudaError_t launch_rbq1_encode(const float *X, int64_t n, int d, const float *m, uint32_t *codes,
+                               float *nx2, float *F, int32_t *popx, cudaStream_t st);
+cudaError_t launch_rbq1_exponent(const float *F, int64_t n, unsigned int *maxbits, int *e_dev,
+                                 cudaStream_t st);
+// centroid preparation
+cudaError_t launch_rbq1_cprep(const float *C, int k, int d, const float *m, uint4 *planes,
+                              Rbq1CInfo *info, cudaStream_t st);
+cudaError_t launch_row_sqnorm_u8(const uint8_t *codes, int64_t n, int d, int32_t *out,
+                                 cudaStream_t st);
+// assignment
+cudaError_t launch_assign_exact_f32(const float *X, int64_t n, int d, const float *C, int k,
+                                    int32_t *assign, float *dist, cudaStream_t st);
+cudaError_t launch_assign_exact_bf16(const uint16_t *X, int64_t n, int d, const float *C, int k,
+                                     int32_t *assign, float *dist, cudaStream_t st);
+cudaError_t launch_assign_sq8_simt(const uint8_t *X, int64_t n, int d, const uint8_t *C, int k,
+                                   const int32_t *nx, const int32_t *nc, int32_t *assign,
+                                   float *dist, cudaStream_t st);
+cudaError_t launch_assign_rbq1(const uint32_t *codes, const float *nx2, const float *F,
+                               const int32_t *popx, int64_t n, int d, const uint4 *planes,
+                               const Rbq1CInfo *info, int k, int32_t *assign, float *dist,
+                               cudaStream_t st);
+// update
+cudaError_t launch_histogram(const int32_t *assign, int64_t n, int k, int32_t *counts32,
+                             cudaStream_t st);
+cudaError_t launch_scan_offsets(const int32_t *counts32, int k, int64_t *offsets,
+                                int64_t *counts64_out, int accumulate_counts, cudaStream_t st);
+cudaError_t launch_scatter(const int32_t *assign, int64_t n, int k, const int64_t *offsets,
+                           int32_t *cursor, int32_t *perm, cudaStream_t st);
+// repr: 0 f32, 3 bf16 (float centroids); mode: 0 finalise, 1 accumulate partial
+cudaError_t launch_segsum_float(const void *X, int x_is_bf16, int d, const int32_t *perm,
+                                const int64_t *offsets, int k, float *C_inout, double *partial,
+                                cudaStream_t st);
+cudaError_t launch_segsum_sq8(const uint8_t *X, int d, const int32_t *perm,
+                              const int64_t *offsets, int k, uint8_t *C_inout, int64_t *partial,
+                              cudaStream_t st);
+cudaError_t launch_segsum_rbq1(const uint32_t *codes, const float *F, int d, const float *m,
+                               int e, const int32_t *perm, const int64_t *offsets, int k,
+                               float *C_inout, int64_t *partial, cudaStream_t st);
+cudaError_t launch_finalize_float(const double *partial, const int64_t *counts, int k, int d,
+                                  float *C_inout, cudaStream_t st);
+cudaError_t launch_finalize_sq8(const int64_t *partial, const int64_t *counts, int k, int d,
+                                uint8_t *C_inout, cudaStream_t st);
+cudaError_t launch_finalize_rbq1(const int64_t *partial, const int64_t *counts, int k, int d,
+                                 const float *m, int e, float *C_inout, cudaStream_t st);
+cudaError_t launch_merge(void *dst, const void *src, int64_t count, int elem_type,
+                         cudaStream_t st);
+// init / objective / projection / pca
+cudaError_t launch_gather_rows(const void *X, int64_t n, int elem_bytes, int64_t row_elems,
+                               const int64_t *idx, int k, void *out, int *status,
+                               cudaStream_t st);
+cudaError_t launch_rbq1_decode_rows(const uint32_t *codes, const float *F, int64_t n, int d,
+                                    const float *m, int e, const int64_t *idx, int k,
+                                    float *out, int *status, cudaStream_t st);
+cudaError_t launch_objective(const void *X, int x_is_bf16, int64_t n, int d, const float *C,
+                             const int32_t *assign, double *partials, int nblk,
+                             cudaStream_t st);
+cudaError_t launch_sum_double(const double *in, int64_t count, double *out, cudaStream_t st);
+cudaError_t launch_sum_float_to_double(const float *in, int64_t count, double *partials,
+                                       int nblk, cudaStream_t st);
+cudaError_t launch_project(const float *X, int64_t n, int d, const float *mean, const float *P,
+                           int d_out, int out_bf16, void *Y, cudaStream_t st);
+cudaError_t launch_cov_partial(const float *X, int64_t n, int d, const float *mean,
+                               double *partial, int splits, cudaStream_t st);
+cudaError_t launch_cov_reduce(const double *partial, int splits, int d, double *cov,
+                              cudaStream_t st);
+
+// host helpers (skm_linalg.cpp)
+void philox_gaussians(uint64_t seed, int64_t count, double *out);
+void householder_qr_q(int d, double *A /* d*d in, Q out, row-major */);
+int symmetric_eigen(int n, double *A /* in: symmetric; out: eigenvectors as columns */,
+                    double *w /* eigenvalues */);
+
+}  // namespace skm

@@ -1,0 +1,97 @@
+"""Host-side checks of the C ABI that need no GPU: the library loads, exports
+every symbol include/skm.h declares, and rejects invalid arguments before
+any launch (so fake device pointers are never dereferenced)."""
+import ctypes
+import os
+import re
+
+import numpy as np
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+@pytest.fixture(scope="module")
+def skm():
+    from paper_2608_14648_gb300 import build as b
+
+    b.build()
+    import paper_2608_14648_gb300 as skm
+
+    return skm
+
+
+def _declared_symbols():
+    src = open(os.path.join(ROOT, "include", "skm.h")).read()
+    return sorted(set(re.findall(r"\b(skm_[a-z0-9_]+)\s*\(", src)))
+
+
+def test_library_exports_every_declared_symbol(skm):
+    declared = _declared_symbols()
+    assert set(declared) == set(skm.EXPORTED_SYMBOLS)
+    L = ctypes.CDLL(skm.lib_path())
+    for name in declared:
+        assert hasattr(L, name), name
+    assert skm.skm_version() >= 100
+
+
+def _data(skm, repr_=0, n=100, d=16):
+    return skm.Data(repr_, d, n, 0x1000, None, None, None, None, 0, 0)
+
+
+FAKE = ctypes.c_void_p(0x1000)
+
+
+def test_invalid_arguments_are_rejected_before_launch(skm):
+    L = skm.lib()
+    x = _data(skm)
+    # k > n
+    rc = L.skm_assign(ctypes.byref(x), FAKE, 101, None, FAKE, None, FAKE, 1 << 20, None)
+    assert rc == 1 and b"exceeds" in L.skm_last_error()
+    # k = 0
+    assert L.skm_assign(ctypes.byref(x), FAKE, 0, None, FAKE, None, FAKE, 1 << 20, None) == 1
+    # d out of range
+    bad = _data(skm, d=0)
+    assert L.skm_assign(ctypes.byref(bad), FAKE, 4, None, FAKE, None, FAKE, 1 << 20, None) == 1
+    big = _data(skm, d=5000)
+    assert L.skm_assign(ctypes.byref(big), FAKE, 4, None, FAKE, None, FAKE, 1 << 20, None) == 2
+    # unknown repr
+    assert L.skm_assign(ctypes.byref(_data(skm, repr_=9)), FAKE, 4, None, FAKE, None, FAKE, 1 << 20, None) == 1
+    # NULL centroids / assign
+    assert L.skm_assign(ctypes.byref(x), None, 4, None, FAKE, None, FAKE, 1 << 20, None) == 1
+    # RBQ1 without its factors
+    r = _data(skm, repr_=2)
+    assert L.skm_assign(ctypes.byref(r), FAKE, 4, None, FAKE, None, FAKE, 1 << 20, None) == 1
+    # workspace too small
+    need = L.skm_workspace_size(0, ctypes.byref(_data(skm, repr_=1)), 4)
+    assert need > 0
+    rc = L.skm_assign(ctypes.byref(_data(skm, repr_=1)), FAKE, 4, None, FAKE, None, FAKE, need - 1, None)
+    assert rc == 4
+    # misaligned workspace
+    rc = L.skm_assign(ctypes.byref(_data(skm, repr_=1)), FAKE, 4, None, FAKE, None, ctypes.c_void_p(0x1010), need,
+                      None)
+    assert rc == 1
+    # fit without any initialisation
+    cfg = skm.FitConfig(4, 3)
+    rc = L.skm_fit(ctypes.byref(cfg), ctypes.byref(x), None, None, FAKE, FAKE, None, None, None, FAKE, 1 << 30, None)
+    assert rc == 1
+    # projection to more dims than the input
+    assert L.skm_project(FAKE, 10, 8, None, FAKE, 9, 0, FAKE, None) == 1
+    # unknown workspace op
+    assert L.skm_workspace_size(7, ctypes.byref(x), 4) == 0
+
+
+def test_workspace_sizes_grow_with_problem(skm):
+    L = skm.lib()
+    small = L.skm_workspace_size(2, ctypes.byref(_data(skm, n=1000, d=64)), 10)
+    large = L.skm_workspace_size(2, ctypes.byref(_data(skm, n=100000, d=64)), 10)
+    assert 0 < small < large
+
+
+def test_make_rotation_is_orthogonal_and_seeded(skm):
+    P = skm.skm_make_rotation(7, 48).numpy().astype(np.float64)
+    np.testing.assert_allclose(P.T @ P, np.eye(48), atol=2e-6)
+    P2 = skm.skm_make_rotation(7, 48).numpy()
+    np.testing.assert_array_equal(P.astype(np.float32), P2)
+    P3 = skm.skm_make_rotation(8, 48).numpy()
+    assert not np.allclose(P2, P3)

@@ -1,0 +1,309 @@
+"""GPU path vs the CPU oracle, element by element, through the C ABI.
+
+Integer paths (SQ8 codes/distances/assignments/centroids, RBQ1 estimates,
+assignments and centroids given identical codes) must be bit-exact; the fp32
+and bf16 paths must agree on >= 99.9% of assignments with every disagreement
+at an oracle top-2 relative gap <= 1e-5, centroids within 1e-4 relative L2
+given identical assignments, objectives within 1e-4 relative."""
+import math
+
+import numpy as np
+import pytest
+import torch
+
+import oracle
+import synth
+
+pytestmark = pytest.mark.gpu
+
+GAP_TOL = 1e-5
+AGREE = 0.999
+
+
+@pytest.fixture(scope="module")
+def skm(cuda_ok):
+    import paper_2608_14648_gb300 as skm
+
+    skm.lib()
+    return skm
+
+
+DEV = "cuda"
+
+
+def _points(n, d, seed, decay=True, ncomp=40):
+    return synth.gmm_points(n, d, ncomp, seed=seed, decay=decay)
+
+
+def _check_f32(a_gpu, dist_gpu, best, second, a_or, what):
+    a_gpu = np.asarray(a_gpu)
+    agree = a_gpu == a_or
+    frac = agree.mean()
+    assert frac >= AGREE, f"{what}: agreement {frac}"
+    if not agree.all():
+        gap = (second - best) / np.maximum(best, 1e-30)
+        assert np.all(gap[~agree] <= GAP_TOL), f"{what}: disagreement at gap {gap[~agree].max()}"
+    if dist_gpu is not None:
+        d = np.asarray(dist_gpu)
+        np.testing.assert_allclose(d[agree], best[agree], rtol=2e-5, atol=1e-6)
+
+
+# ----------------------------------------------------------------- fp32 path
+@pytest.mark.parametrize("n,d,k", [(1000, 128, 100), (777, 33, 7), (3001, 768, 300), (200, 1, 5),
+                                   (513, 64, 257), (64, 200, 64)])
+def test_assign_f32_vs_oracle(skm, n, d, k):
+    X = _points(n, d, seed=n + d)
+    idx = synth.forgy_indices(n, k, seed=d)
+    C = X[idx].clone()
+    C += 0.01 * torch.randn(C.shape, generator=torch.Generator().manual_seed(1))
+    pts = skm.Points(skm.REPR_F32, X.to(DEV), d)
+    a, dist = skm.skm_assign(pts, C.to(DEV))
+    a_or, best, second = oracle.assign_f32(X.numpy(), C.numpy())
+    _check_f32(a.cpu().numpy(), dist.cpu().numpy(), best, second, a_or, f"f32 n={n} d={d} k={k}")
+
+
+def test_assign_f32_edge_cases(skm):
+    X = _points(300, 40, seed=3)
+    Xd = X.to(DEV)
+    pts = skm.Points(skm.REPR_F32, Xd, 40)
+    # k = 1
+    a, _ = skm.skm_assign(pts, Xd[:1].clone())
+    assert torch.all(a == 0)
+    # n = k with centroids = points: identity, zero distance
+    a, dist = skm.skm_assign(pts, Xd.clone())
+    assert torch.equal(a.cpu(), torch.arange(300, dtype=torch.int32))
+    assert float(dist.abs().max()) == 0.0
+    # duplicated centroids: ties go to the lowest index
+    C = torch.cat([Xd[5:6], Xd[5:6], Xd[9:10], Xd[9:10]]).contiguous()
+    sub = skm.Points(skm.REPR_F32, Xd[[5, 9]].contiguous(), 40)
+    a, _ = skm.skm_assign(sub, C)
+    assert a.tolist() == [0, 2]
+
+
+def test_update_f32_vs_oracle(skm):
+    n, d, k = 5000, 100, 37
+    X = _points(n, d, seed=4)
+    a = torch.randint(0, k - 1, (n,), generator=torch.Generator().manual_seed(2), dtype=torch.int32)
+    C0 = torch.randn(k, d, generator=torch.Generator().manual_seed(3))
+    pts = skm.Points(skm.REPR_F32, X.to(DEV), d)
+    C, counts = skm.skm_update(pts, a.to(DEV), C0.to(DEV).clone())
+    Co, co = oracle.update_f32(X.numpy(), a.numpy(), C0.numpy())
+    np.testing.assert_array_equal(counts.cpu().numpy(), co)
+    Cg = C.cpu().numpy().astype(np.float64)
+    rel = np.linalg.norm(Cg - Co, axis=1) / np.maximum(np.linalg.norm(Co, axis=1), 1e-30)
+    assert rel.max() <= 1e-4
+    np.testing.assert_array_equal(C.cpu().numpy()[k - 1], C0.numpy()[k - 1])  # empty cluster kept
+
+
+def test_fit_f32_tiny_workload(skm):
+    spec = synth.WORKLOADS["tiny_f32"]
+    X = synth.workload_points(spec, seed=0)
+    idx = synth.forgy_indices(spec.n, spec.k, seed=0)
+    pts = skm.Points(skm.REPR_F32, X.to(DEV), spec.d)
+    C, a, dist, obj, stats = skm.skm_fit(pts, spec.k, spec.iters, init_idx=idx.to(DEV))
+    Co, ao, objo = oracle.lloyd_f32(X.numpy(), X.numpy()[idx.numpy()], spec.iters)
+    agree = (a.cpu().numpy() == ao).mean()
+    assert agree >= AGREE
+    assert abs(obj[-1] - objo[-1]) / objo[-1] <= 1e-4
+    # the GPU trajectory's objective is non-increasing too
+    for t in range(1, len(obj)):
+        assert obj[t] <= obj[t - 1] * (1 + 1e-6)
+    # final objective recomputed in fp64 from the GPU's own outputs
+    full = oracle.objective_f32(X.numpy(), C.cpu().numpy(), a.cpu().numpy())
+    assert abs(full - objo[-1]) / objo[-1] <= 1e-4
+
+
+# ------------------------------------------------------------------ SQ8 path
+@pytest.mark.parametrize("n,d", [(2000, 64), (777, 33), (1500, 1024), (50, 1)])
+def test_quantize_sq8_bitexact(skm, n, d):
+    X = _points(n, d, seed=n)
+    q = skm.skm_quantize(skm.REPR_SQ8, X.to(DEV))
+    b, s = oracle.sq8_fit(X.numpy())
+    np.testing.assert_array_equal(q["b"].cpu().numpy(), b)
+    np.testing.assert_array_equal(q["s"].cpu().numpy(), s)
+    np.testing.assert_array_equal(q["codes"].cpu().numpy(), oracle.sq8_encode(X.numpy(), b, s))
+    Y = skm.skm_sq8_decode(q["codes"], q["b"], q["s"])
+    np.testing.assert_array_equal(Y.cpu().numpy(), oracle.sq8_decode(q["codes"].cpu().numpy(), b, s))
+
+
+@pytest.mark.parametrize("n,d,k", [(2000, 64, 50), (777, 33, 7), (1024, 1024, 129), (300, 5, 300)])
+def test_assign_update_sq8_bitexact(skm, n, d, k):
+    g = np.random.default_rng(n + d)
+    Xc = g.integers(0, 256, size=(n, d)).astype(np.uint8)
+    Cc = Xc[g.choice(n, k, replace=False)].copy()
+    if k > 3:
+        Cc[3] = Cc[1]  # duplicate
+    pts = skm.Points(skm.REPR_SQ8, torch.from_numpy(Xc).to(DEV), d)
+    a, dist = skm.skm_assign(pts, torch.from_numpy(Cc).to(DEV))
+    ao, bo = oracle.assign_sq8(Xc, Cc)
+    np.testing.assert_array_equal(a.cpu().numpy(), ao)
+    np.testing.assert_array_equal(dist.cpu().numpy(), bo.astype(np.float32))
+    C, counts = skm.skm_update(pts, a, torch.from_numpy(Cc).to(DEV).clone())
+    Co, co = oracle.update_sq8(Xc, ao, Cc)
+    np.testing.assert_array_equal(counts.cpu().numpy(), co)
+    np.testing.assert_array_equal(C.cpu().numpy(), Co)
+
+
+def test_fit_sq8_trajectory_bitexact(skm):
+    n, d, k, iters = 6000, 256, 64, 6
+    X = _points(n, d, seed=8)
+    q = skm.skm_quantize(skm.REPR_SQ8, X.to(DEV))
+    idx = synth.forgy_indices(n, k, seed=8)
+    C, a, _, _, _ = skm.skm_fit(skm.Points(skm.REPR_SQ8, q["codes"], d), k, iters, init_idx=idx.to(DEV))
+    codes = q["codes"].cpu().numpy()
+    Co, ao = oracle.lloyd_sq8(codes, codes[idx.numpy()], iters)
+    np.testing.assert_array_equal(a.cpu().numpy(), ao)
+    np.testing.assert_array_equal(C.cpu().numpy(), Co)
+
+
+# ---------------------------------------------------------------- RBQ1 path
+def _rbq1_host(r):
+    h = {k: v.cpu().numpy() for k, v in r.items()}
+    h["codes"] = h["codes"].view(np.uint32)
+    return h
+
+
+@pytest.mark.parametrize("n,d", [(3000, 768), (777, 33), (500, 32), (400, 31), (100, 1)])
+def test_encode_rbq1_vs_oracle(skm, n, d):
+    X = _points(n, d, seed=n + 1)
+    r = skm.skm_quantize(skm.REPR_RBQ1, X.to(DEV))
+    h = _rbq1_host(r)
+    m = oracle.rbq1_mean(X.numpy())
+    np.testing.assert_allclose(h["m"], m, rtol=1e-6, atol=1e-7)
+    # codes from the GPU's own mean must match the oracle's encoder bit for bit
+    codes, nx2, F, popx = oracle.rbq1_encode(X.numpy(), h["m"])
+    np.testing.assert_array_equal(h["codes"], codes)
+    np.testing.assert_array_equal(h["popx"], popx)
+    np.testing.assert_allclose(h["nx2"], nx2, rtol=1e-6)
+    np.testing.assert_allclose(h["F"], F, rtol=1e-6)
+    # unused high bits of the last word are zero
+    if d % 32:
+        assert np.all(h["codes"][:, -1] >> (d % 32) == 0)
+
+
+@pytest.mark.parametrize("n,d,k", [(3000, 768, 300), (777, 33, 7), (500, 64, 1), (1000, 1024, 65)])
+def test_assign_update_rbq1_bitexact(skm, n, d, k):
+    X = _points(n, d, seed=n + 2)
+    r = skm.skm_quantize(skm.REPR_RBQ1, X.to(DEV))
+    pts = skm.rbq1_points(r, d)
+    h = _rbq1_host(r)
+    assert pts.rbq1_exp == oracle.rbq1_exponent(h["F"])
+    C = X[synth.forgy_indices(n, k, seed=5)].clone()
+    a, est = skm.skm_assign(pts, C.to(DEV))
+    prep = oracle.rbq1_centroid_sq4(C.numpy(), h["m"])
+    ao, esto = oracle.rbq1_assign(h["codes"], h["nx2"], h["F"], h["popx"], d, prep)
+    np.testing.assert_array_equal(a.cpu().numpy(), ao)
+    np.testing.assert_array_equal(est.cpu().numpy(), esto)
+    Cn, counts = skm.skm_update(pts, a, C.to(DEV).clone())
+    Co, co = oracle.rbq1_update(h["codes"], h["F"], d, h["m"], pts.rbq1_exp, ao, C.numpy())
+    np.testing.assert_array_equal(counts.cpu().numpy(), co)
+    np.testing.assert_array_equal(Cn.cpu().numpy(), Co)
+
+
+def test_fit_rbq1_trajectory_bitexact(skm):
+    n, d, k, iters = 8000, 256, 50, 6
+    X = _points(n, d, seed=9)
+    r = skm.skm_quantize(skm.REPR_RBQ1, X.to(DEV))
+    pts = skm.rbq1_points(r, d)
+    idx = synth.forgy_indices(n, k, seed=9)
+    C, a, _, _, _ = skm.skm_fit(pts, k, iters, init_idx=idx.to(DEV))
+    h = _rbq1_host(r)
+    C0 = oracle.rbq1_decode_points(h["codes"], h["F"], d, h["m"], pts.rbq1_exp, idx.numpy())
+    Co, ao = oracle.lloyd_rbq1(h["codes"], h["nx2"], h["F"], h["popx"], d, h["m"], C0, iters, pts.rbq1_exp)
+    np.testing.assert_array_equal(a.cpu().numpy(), ao)
+    np.testing.assert_array_equal(C.cpu().numpy(), Co)
+
+
+# ------------------------------------------------------ projection and bf16
+@pytest.mark.parametrize("n,d,dout", [(1000, 128, 128), (777, 100, 33), (2048, 1024, 256)])
+def test_project_vs_oracle(skm, n, d, dout):
+    X = _points(n, d, seed=d)
+    P = synth.haar_rotation(d, 4)[:, :dout].to(torch.float32).contiguous()
+    mu = X.mean(0)
+    Y = skm.skm_project(X.to(DEV), P.to(DEV), mu.to(DEV))
+    Yo = oracle.project(X.numpy(), P.numpy(), mu.numpy())
+    scale = np.linalg.norm(X.numpy() - mu.numpy(), axis=1)[:, None]
+    assert np.max(np.abs(Y.cpu().numpy() - Yo) / scale) < 2e-6
+    Yb = skm.skm_project(X.to(DEV), P.to(DEV), mu.to(DEV), out_dtype=skm.DTYPE_BF16)
+    yb = Yb.view(torch.int16).cpu().numpy().view(np.uint16)
+    ybo = oracle.round_bf16(Yo)
+    # bf16 of the fp32 result vs bf16 of the fp64 result: equal or 1 ulp apart
+    diff = np.abs(yb.astype(np.int32) - ybo.astype(np.int32))
+    assert diff.max() <= 1 and (diff == 0).mean() > 0.99
+
+
+@pytest.mark.parametrize("n,d,k", [(2000, 256, 100), (777, 64, 13), (300, 32, 300)])
+def test_assign_update_bf16_vs_oracle(skm, n, d, k):
+    X = _points(n, d, seed=n)
+    Xb = X.to(DEV).to(torch.bfloat16)
+    xb = Xb.view(torch.int16).cpu().numpy().view(np.uint16)
+    C = oracle.bf16_to_f32(xb[synth.forgy_indices(n, k, seed=3).numpy()]).copy()
+    pts = skm.Points(skm.REPR_BF16, Xb.view(torch.int16), d)
+    a, dist = skm.skm_assign(pts, torch.from_numpy(C).to(DEV))
+    a_or, best, second = oracle.assign_bf16(xb, C)
+    _check_f32(a.cpu().numpy(), dist.cpu().numpy(), best, second, a_or, "bf16")
+    Cn, counts = skm.skm_update(pts, torch.from_numpy(a_or).to(DEV), torch.from_numpy(C).to(DEV).clone())
+    Co, co = oracle.update_bf16(xb, a_or, C)
+    np.testing.assert_array_equal(counts.cpu().numpy(), co)
+    rel = np.linalg.norm(Cn.cpu().numpy() - Co, axis=1) / np.maximum(np.linalg.norm(Co, axis=1), 1e-30)
+    assert rel.max() <= 1e-4
+
+
+def test_pca_fit_vs_oracle(skm):
+    n, d, dout = 20000, 64, 16
+    X = _points(n, d, seed=12)
+    mean, P, w = skm.skm_pca_fit(X.to(DEV), dout)
+    mu, Po, wo = oracle.pca_fit(X.numpy(), dout)
+    np.testing.assert_allclose(mean.cpu().numpy(), mu, rtol=1e-5, atol=1e-7)
+    np.testing.assert_allclose(w.cpu().numpy(), wo, rtol=1e-4)
+    # eigenvectors agree where the spectrum is separated (sign fixed on both sides)
+    gaps = np.abs(np.diff(np.concatenate([wo, [0.0]]))) / wo
+    sep = gaps > 1e-2
+    sep[1:] &= gaps[:-1] > 1e-2
+    Pg = P.cpu().numpy()
+    for j in np.where(sep)[0]:
+        assert abs(float(Pg[:, j] @ Po[:, j])) > 0.999
+
+
+# --------------------------------------------------------- sharded update
+@pytest.mark.parametrize("repr_name", ["f32", "sq8", "rbq1"])
+def test_sharded_update_matches_single(skm, repr_name):
+    n, d, k = 4000, 64, 20
+    X = _points(n, d, seed=21)
+    Xd = X.to(DEV)
+    if repr_name == "f32":
+        pts = skm.Points(skm.REPR_F32, Xd, d)
+        C = Xd[:k].clone()
+        pdt, pshape = torch.float64, (k, d)
+    elif repr_name == "sq8":
+        q = skm.skm_quantize(skm.REPR_SQ8, Xd)
+        pts = skm.Points(skm.REPR_SQ8, q["codes"], d)
+        C = q["codes"][:k].clone()
+        pdt, pshape = torch.int64, (k, d)
+    else:
+        r = skm.skm_quantize(skm.REPR_RBQ1, Xd)
+        pts = skm.rbq1_points(r, d)
+        C = Xd[:k].clone()
+        pdt, pshape = torch.int64, (k, d + 1)
+    a, _ = skm.skm_assign(pts, C)
+    C_single, cnt_single = skm.skm_update(pts, a, C.clone())
+    bounds = [0, 1000, 1001, 2777, n]
+    total = torch.zeros(pshape, dtype=pdt, device=DEV)
+    counts = torch.zeros(k, dtype=torch.int64, device=DEV)
+    for lo, hi in zip(bounds[:-1], bounds[1:]):
+        part = torch.zeros(pshape, dtype=pdt, device=DEV)
+        sub_x = pts.x[lo:hi].contiguous()
+        extra = {}
+        if repr_name == "rbq1":
+            extra = dict(nx2=pts.nx2[lo:hi].contiguous(), F=pts.F[lo:hi].contiguous(),
+                         popx=pts.popx[lo:hi].contiguous(), m=pts.m, rbq1_exp=pts.rbq1_exp)
+        sp = skm.Points(pts.repr, sub_x, d, **extra)
+        skm.skm_update(sp, a[lo:hi].contiguous(), None, counts=counts, partial=part)
+        skm.skm_merge_partials(total, part)
+    C_merged = skm.skm_update_finalize(pts, total, counts, C.clone())
+    assert torch.equal(counts, cnt_single)
+    if repr_name == "f32":
+        rel = (C_merged - C_single).norm(dim=1) / C_single.norm(dim=1)
+        assert float(rel.max()) <= 1e-5
+    else:
+        assert torch.equal(C_merged, C_single)
