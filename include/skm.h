@@ -73,6 +73,10 @@ typedef struct skm_data {
     int32_t rbq1_exp;   /* fixed-point exponent e of the decode-average
                            (skm_rbq1_exponent); fit() computes it itself     */
     int32_t reserved0;
+    /* Optional screening copy for F32 / BF16 / SQ8 assignment, built once by
+     * skm_screen_prep (the points never change across Lloyd iterations).
+     * NULL: skm_assign builds it in its workspace on every call.            */
+    const void *screen;
 } skm_data;
 
 /* Optional per-call statistics (host struct, filled after the call's work
@@ -162,6 +166,16 @@ int skm_quantize(int repr, const float *X, int64_t n, int d, skm_quant_params *q
 int skm_rbq1_exponent(const float *F, int64_t n, int *e_host, void *ws, size_t ws_bytes,
                       void *stream);
 
+/* Screening copy of the points for the tensor-core assignment (opaque
+ * layout): F32 -> bf16 copy + per-point (||x~||, ||x~ - x||); SQ8 -> centred
+ * codes (code - 128) in bf16 + centred squared norms; BF16 -> per-point norms
+ * (plus a padded copy when d is not a multiple of 8).  skm_screen_bytes
+ * returns its size (0 when the representation needs none: RBQ1, or SQ8 with
+ * d > 1024); skm_screen_prep fills `screen` (device, 256-byte aligned,
+ * caller-owned) from x->x.  Asynchronous. */
+size_t skm_screen_bytes(const skm_data *x);
+int skm_screen_prep(const skm_data *x, void *screen, size_t screen_bytes, void *stream);
+
 /* ------------------------------------------------------------------------
  * Assignment, Section 2.3 STEP 2: assign[p] = argmin_j dist(x_p, c_j).
  *  C (device), per repr:
@@ -199,6 +213,7 @@ int skm_assign(const skm_data *x, const void *C, int k, const int32_t *prev_assi
  *             / count_j) / sqrt(d) in fp64, rounded to fp32, where
  *             T_ji = sum Fq xbar_i, U_j = sum Fq, Fq = round(F 2^e) (int64,
  *             exact), e = x->rbq1_exp.
+ *  Assignments outside [0, k) are skipped (not counted, not summed).
  *  partial != NULL selects the sharded form: nothing is finalised; the
  *  cluster sums are ADDED into `partial` and the member counts into
  *  `counts` (both zeroed by the caller before the first shard) so that
@@ -224,6 +239,9 @@ int skm_update_finalize(const skm_data *x, const void *partial, const int64_t *c
  *  skm_assign) when non-NULL, else the points init_idx[0..k) (device int64,
  *  Forgy, STEP 1): F32/BF16 rows, SQ8 codes, RBQ1 decoded points (the
  *  decode-average of one member).
+ *  An init_idx entry outside [0, n) makes the call fail with
+ *  SKM_ERR_DEVICE_CHECK before any iteration; a tensor-core pipeline wait
+ *  that exceeds its 2 s limit makes it return SKM_ERR_TIMEOUT.
  *  Outputs (device): C_out (per-repr layout), assign_out int32[n],
  *  dist_out float[n] or NULL (from the final assignment).
  *  objective_host (host, iters+1 doubles, may be NULL): sum of the

@@ -30,7 +30,8 @@ _lib = None
 
 # Every entry point declared in include/skm.h.
 EXPORTED_SYMBOLS = [
-    "skm_last_error", "skm_version", "skm_kernel_launches", "skm_workspace_size", "skm_project", "skm_make_rotation",
+    "skm_last_error", "skm_version", "skm_kernel_launches", "skm_workspace_size", "skm_screen_bytes",
+    "skm_screen_prep", "skm_project", "skm_make_rotation",
     "skm_pca_fit", "skm_quantize", "skm_rbq1_exponent", "skm_assign", "skm_update",
     "skm_merge_partials", "skm_update_finalize", "skm_fit", "skm_objective", "skm_sq8_decode",
 ]
@@ -49,7 +50,7 @@ class Data(ctypes.Structure):
         ("repr", ctypes.c_int32), ("d", ctypes.c_int32), ("n", ctypes.c_int64),
         ("x", ctypes.c_void_p), ("nx2", ctypes.c_void_p), ("F", ctypes.c_void_p),
         ("popx", ctypes.c_void_p), ("m", ctypes.c_void_p), ("rbq1_exp", ctypes.c_int32),
-        ("reserved0", ctypes.c_int32),
+        ("reserved0", ctypes.c_int32), ("screen", ctypes.c_void_p),
     ]
 
 
@@ -87,6 +88,8 @@ def lib():
             "skm_version": ([], i32),
             "skm_kernel_launches": ([], ctypes.c_uint64),
             "skm_workspace_size": ([i32, vp, i32], sz),
+            "skm_screen_bytes": ([vp], sz),
+            "skm_screen_prep": ([vp, vp, sz, vp], i32),
             "skm_project": ([vp, i64, i32, vp, vp, i32, i32, vp, vp], i32),
             "skm_make_rotation": ([u64, i32, vp], i32),
             "skm_pca_fit": ([vp, i64, i32, i32, vp, vp, vp, vp, sz, vp], i32),
@@ -135,14 +138,24 @@ def _dev(t):
 class Points:
     """Keeps the tensors of one skm_data alive; `.ref` is the ctypes struct."""
 
-    def __init__(self, repr_, x, d, nx2=None, F=None, popx=None, m=None, rbq1_exp=0):
+    def __init__(self, repr_, x, d, nx2=None, F=None, popx=None, m=None, rbq1_exp=0, screen=None):
         assert x.is_contiguous()
         self.repr, self.x, self.d = repr_, x, int(d)
         self.nx2, self.F, self.popx, self.m = nx2, F, popx, m
         self.n = x.shape[0]
         self.rbq1_exp = int(rbq1_exp)
+        self.screen = screen
         self.ref = Data(repr_, self.d, self.n, x.data_ptr(), _ptr(nx2), _ptr(F), _ptr(popx), _ptr(m),
-                        self.rbq1_exp, 0)
+                        self.rbq1_exp, 0, _ptr(screen))
+
+    def with_screen(self, stream=None):
+        """Builds the screening copy once (skm_screen_prep) and attaches it."""
+        nbytes = lib().skm_screen_bytes(ctypes.byref(self.ref))
+        if nbytes == 0:
+            return self
+        buf = _ws(nbytes, self.device)
+        _check(lib().skm_screen_prep(ctypes.byref(self.ref), _ptr(buf), buf.numel(), _stream(stream)))
+        return Points(self.repr, self.x, self.d, self.nx2, self.F, self.popx, self.m, self.rbq1_exp, buf)
 
     @property
     def device(self):

@@ -30,10 +30,14 @@ __device__ __forceinline__ void argmin_merge(float &bd, int &bi, float d, int i)
     }
 }
 
+// rows == nullptr: rows 0..nrows-1.  Otherwise the rows are rows[0..count)
+// with count = *nrows_dev (a device-side list, e.g. the rows a screen could
+// not decide).  Blocks stride over 64-row tiles.
 template <typename TX>
 __global__ void __launch_bounds__(256) assign_exact_kernel(const TX *__restrict__ X,
                                                            const int32_t *__restrict__ rows,
-                                                           int64_t nrows, int d,
+                                                           const int32_t *__restrict__ nrows_dev,
+                                                           int64_t nrows_arg, int d,
                                                            const float *__restrict__ C, int k,
                                                            int32_t *__restrict__ assign,
                                                            float *__restrict__ dist) {
@@ -41,117 +45,139 @@ __global__ void __launch_bounds__(256) assign_exact_kernel(const TX *__restrict_
     __shared__ __align__(16) float cs[32][68];
     const int tid = threadIdx.x;
     const int ty = tid >> 4, tx = tid & 15;
-    const int64_t row0 = (int64_t)blockIdx.x * 64;
+    const int64_t nrows = nrows_dev ? (int64_t)*nrows_dev : nrows_arg;
+    for (int64_t row0 = (int64_t)blockIdx.x * 64; row0 < nrows; row0 += (int64_t)gridDim.x * 64) {
+        __syncthreads();
 
-    // the point rows this block owns (indirect when `rows` is given)
-    int64_t prow[4];
-    bool pval[4];
-#pragma unroll
-    for (int i = 0; i < 4; ++i) {
-        const int64_t r = row0 + ty * 4 + i;
-        pval[i] = r < nrows;
-        prow[i] = pval[i] ? (rows ? (int64_t)rows[r] : r) : 0;
-    }
-    // loader mapping: thread loads rows lr0 + 8q (q = 0..7) at dim ld
-    const int ld = tid & 31, lr0 = tid >> 5;
-    int64_t lrow[8];
-    bool lval[8];
-#pragma unroll
-    for (int q = 0; q < 8; ++q) {
-        const int64_t r = row0 + lr0 + 8 * q;
-        lval[q] = r < nrows;
-        lrow[q] = lval[q] ? (rows ? (int64_t)rows[r] : r) : 0;
-    }
-
-    float best[4];
-    int besti[4];
-#pragma unroll
-    for (int i = 0; i < 4; ++i) {
-        best[i] = INFINITY;
-        besti[i] = 0x7fffffff;
-    }
-
-    for (int c0 = 0; c0 < k; c0 += 64) {
-        float acc[4][4];
-#pragma unroll
-        for (int i = 0; i < 4; ++i)
-#pragma unroll
-            for (int j = 0; j < 4; ++j) acc[i][j] = 0.0f;
-
-        for (int k0 = 0; k0 < d; k0 += 32) {
-            const int dim = k0 + ld;
-            __syncthreads();
-#pragma unroll
-            for (int q = 0; q < 8; ++q) {
-                const int r = lr0 + 8 * q;
-                float xv = 0.0f, cv = 0.0f;
-                if (dim < d) {
-                    if (lval[q]) xv = load_x<TX>(X + lrow[q] * d + dim);
-                    if (c0 + r < k) cv = __ldg(C + (int64_t)(c0 + r) * d + dim);
-                }
-                xs[ld][r] = xv;
-                cs[ld][r] = cv;
-            }
-            __syncthreads();
-            const int kmax = min(32, d - k0);
-            for (int kk = 0; kk < kmax; ++kk) {
-                const float4 xv = *reinterpret_cast<const float4 *>(&xs[kk][ty * 4]);
-                const float4 cv = *reinterpret_cast<const float4 *>(&cs[kk][tx * 4]);
-                const float xa[4] = {xv.x, xv.y, xv.z, xv.w};
-                const float ca[4] = {cv.x, cv.y, cv.z, cv.w};
-#pragma unroll
-                for (int i = 0; i < 4; ++i)
-#pragma unroll
-                    for (int j = 0; j < 4; ++j) {
-                        const float t = __fsub_rn(xa[i], ca[j]);
-                        acc[i][j] = __fmaf_rn(t, t, acc[i][j]);
-                    }
-            }
-        }
-        // per-row argmin over this centroid tile, then merge into the running best
+        // the point rows this block owns (indirect when `rows` is given)
+        int64_t prow[4];
+        bool pval[4];
 #pragma unroll
         for (int i = 0; i < 4; ++i) {
-            float bd = INFINITY;
-            int bi = 0x7fffffff;
-#pragma unroll
-            for (int j = 0; j < 4; ++j) {
-                const int cj = c0 + tx * 4 + j;
-                if (cj < k) argmin_merge(bd, bi, acc[i][j], cj);
-            }
-#pragma unroll
-            for (int o = 8; o > 0; o >>= 1) {
-                const float od = __shfl_xor_sync(0xffffffffu, bd, o);
-                const int oi = __shfl_xor_sync(0xffffffffu, bi, o);
-                argmin_merge(bd, bi, od, oi);
-            }
-            argmin_merge(best[i], besti[i], bd, bi);
+            const int64_t r = row0 + ty * 4 + i;
+            pval[i] = r < nrows;
+            prow[i] = pval[i] ? (rows ? (int64_t)rows[r] : r) : 0;
         }
-    }
-    if (tx == 0) {
+        // loader mapping: thread loads rows lr0 + 8q (q = 0..7) at dim ld
+        const int ld = tid & 31, lr0 = tid >> 5;
+        int64_t lrow[8];
+        bool lval[8];
 #pragma unroll
-        for (int i = 0; i < 4; ++i)
-            if (pval[i]) {
-                assign[prow[i]] = besti[i];
-                if (dist) dist[prow[i]] = best[i];
+        for (int q = 0; q < 8; ++q) {
+            const int64_t r = row0 + lr0 + 8 * q;
+            lval[q] = r < nrows;
+            lrow[q] = lval[q] ? (rows ? (int64_t)rows[r] : r) : 0;
+        }
+
+        float best[4];
+        int besti[4];
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+            best[i] = INFINITY;
+            besti[i] = 0x7fffffff;
+        }
+
+        for (int c0 = 0; c0 < k; c0 += 64) {
+            float acc[4][4];
+#pragma unroll
+            for (int i = 0; i < 4; ++i)
+#pragma unroll
+                for (int j = 0; j < 4; ++j) acc[i][j] = 0.0f;
+
+            for (int k0 = 0; k0 < d; k0 += 32) {
+                const int dim = k0 + ld;
+                __syncthreads();
+#pragma unroll
+                for (int q = 0; q < 8; ++q) {
+                    const int r = lr0 + 8 * q;
+                    float xv = 0.0f, cv = 0.0f;
+                    if (dim < d) {
+                        if (lval[q]) xv = load_x<TX>(X + lrow[q] * d + dim);
+                        if (c0 + r < k) cv = __ldg(C + (int64_t)(c0 + r) * d + dim);
+                    }
+                    xs[ld][r] = xv;
+                    cs[ld][r] = cv;
+                }
+                __syncthreads();
+                const int kmax = min(32, d - k0);
+                for (int kk = 0; kk < kmax; ++kk) {
+                    const float4 xv = *reinterpret_cast<const float4 *>(&xs[kk][ty * 4]);
+                    const float4 cv = *reinterpret_cast<const float4 *>(&cs[kk][tx * 4]);
+                    const float xa[4] = {xv.x, xv.y, xv.z, xv.w};
+                    const float ca[4] = {cv.x, cv.y, cv.z, cv.w};
+#pragma unroll
+                    for (int i = 0; i < 4; ++i)
+#pragma unroll
+                        for (int j = 0; j < 4; ++j) {
+                            const float t = __fsub_rn(xa[i], ca[j]);
+                            acc[i][j] = __fmaf_rn(t, t, acc[i][j]);
+                        }
+                }
             }
-    }
+            // per-row argmin over this centroid tile, then merge into the running best
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+                float bd = INFINITY;
+                int bi = 0x7fffffff;
+#pragma unroll
+                for (int j = 0; j < 4; ++j) {
+                    const int cj = c0 + tx * 4 + j;
+                    if (cj < k) argmin_merge(bd, bi, acc[i][j], cj);
+                }
+#pragma unroll
+                for (int o = 8; o > 0; o >>= 1) {
+                    const float od = __shfl_xor_sync(0xffffffffu, bd, o);
+                    const int oi = __shfl_xor_sync(0xffffffffu, bi, o);
+                    argmin_merge(bd, bi, od, oi);
+                }
+                argmin_merge(best[i], besti[i], bd, bi);
+            }
+        }
+        if (tx == 0) {
+#pragma unroll
+            for (int i = 0; i < 4; ++i)
+                if (pval[i]) {
+                    assign[prow[i]] = besti[i];
+                    if (dist) dist[prow[i]] = best[i];
+                }
+        }
+    }  // row tiles
 }
 
-static unsigned blocks_for_rows(int64_t nrows) { return (unsigned)((nrows + 63) / 64); }
+static unsigned blocks_for_rows(int64_t nrows) {
+    int64_t b = (nrows + 63) / 64;
+    const int64_t cap = 152LL * 8;  // 8 resident 256-thread blocks per SM
+    return (unsigned)(b < 1 ? 1 : (b > cap ? cap : b));
+}
 
 cudaError_t launch_assign_exact_f32(const float *X, int64_t n, int d, const float *C, int k,
                                     int32_t *assign, float *dist, cudaStream_t st) {
     if (n == 0) return cudaSuccess;
-    assign_exact_kernel<float><<<blocks_for_rows(n), 256, 0, st>>>(X, nullptr, n, d, C, k,
-                                                                   assign, dist);
+    assign_exact_kernel<float><<<blocks_for_rows(n), 256, 0, st>>>(X, nullptr, nullptr, n, d, C,
+                                                                   k, assign, dist);
     return launched();
 }
 
 cudaError_t launch_assign_exact_bf16(const uint16_t *X, int64_t n, int d, const float *C, int k,
                                      int32_t *assign, float *dist, cudaStream_t st) {
     if (n == 0) return cudaSuccess;
-    assign_exact_kernel<uint16_t><<<blocks_for_rows(n), 256, 0, st>>>(X, nullptr, n, d, C, k,
-                                                                      assign, dist);
+    assign_exact_kernel<uint16_t><<<blocks_for_rows(n), 256, 0, st>>>(X, nullptr, nullptr, n, d,
+                                                                      C, k, assign, dist);
+    return launched();
+}
+
+cudaError_t launch_assign_exact_rows(const void *X, int x_is_bf16, const int32_t *rows,
+                                     const int32_t *count_dev, int64_t max_rows, int d,
+                                     const float *C, int k, int32_t *assign, float *dist,
+                                     cudaStream_t st) {
+    if (max_rows == 0) return cudaSuccess;
+    const unsigned g = blocks_for_rows(max_rows);
+    if (x_is_bf16)
+        assign_exact_kernel<uint16_t><<<g, 256, 0, st>>>(static_cast<const uint16_t *>(X), rows,
+                                                         count_dev, 0, d, C, k, assign, dist);
+    else
+        assign_exact_kernel<float><<<g, 256, 0, st>>>(static_cast<const float *>(X), rows,
+                                                      count_dev, 0, d, C, k, assign, dist);
     return launched();
 }
 

@@ -1,36 +1,882 @@
-// Assignment for the dense representations.
+// Tensor-core assignment (Section 2.3 STEP 2 "GEMM of the data points and
+// centroids", Section 3.1 8-bit GEMM) on sm_103a with tcgen05 + TMEM + TMA.
+//
+// One persistent CTA per SM walks (point tile, centroid tile) jobs:
+//   warp 0      TMA producer: 128 x 64 point slice and 256 x 64 centroid slice
+//               (bf16, 128-byte swizzle) per stage, 4-stage mbarrier ring
+//   warp 1      MMA issuer: 4 x tcgen05.mma.kind::f16 (M=128, N=256, K=16)
+//               per stage into one of two 128 x 256 fp32 TMEM accumulators
+//   warps 2-5   epilogue: tcgen05.ld of the accumulator (thread = point row),
+//               fused per-row reduction over centroids, so the N x K distance
+//               matrix never leaves the SM
+// Two epilogues:
+//  SCREEN (fp32 / bf16 points): bf16 operands, so the dot product carries a
+//    rounding error.  Each pair gets a rigorous interval [L, U] for
+//    s = ||c||^2 - 2 x.c (the distance minus ||x||^2) from per-row and
+//    per-centroid bf16 residual norms.  Per row the epilogue keeps the T
+//    smallest L, the smallest U (Umin) and the smallest L it did not keep
+//    (Lev).  The nearest centroid has L <= Umin, so a row whose only such
+//    candidate is its first is decided; rows with 2..T candidates are
+//    re-scored exactly in fp32; rows with Lev <= Umin are rescanned over all
+//    k in fp32.
+//  SQ8: centred codes (code - 128) are exact in bf16 and every partial sum is
+//    an integer below 2^24 for d <= 1024, so the fp32 accumulator holds the
+//    exact integer dot product; the epilogue forms the integer distance and
+//    keeps the argmin (ties to the lowest index).
+#include <cuda.h>
+#include <cudaTypedefs.h>
+
+#include <mutex>
+
 #include "skm_tc.cuh"
 
 namespace skm {
+namespace {
 
-void tc_plan(int repr, int64_t n, int d, int k, Carver &cv, TcAssignBufs &b) {
-    (void)repr; (void)n; (void)d; (void)k;
-    b.stats = cv.take<int64_t>(2);
+constexpr int BM = 128;  // points per tile (TMEM lanes)
+constexpr int BN = 256;  // centroids per tile (fp32 accumulator columns)
+constexpr int BK = 64;   // bf16 elements per 128-byte swizzle row
+constexpr int STAGES = 4;
+constexpr int A_STAGE = BM * BK * 2;  // 16 KiB
+constexpr int B_STAGE = BN * BK * 2;  // 32 KiB
+constexpr int EPI_WARPS = 4;
+constexpr int THREADS = 64 + 32 * EPI_WARPS;
+constexpr int TCAND = 4;
+constexpr unsigned long long WAIT_LIMIT_NS = 2000000000ull;  // 2 s per barrier wait
+constexpr size_t SMEM_BYTES = 1024 + (size_t)STAGES * (A_STAGE + B_STAGE) + 256;
+
+enum { MODE_SCREEN = 0, MODE_SQ8 = 1 };
+
+struct TcParams {
+    int64_t n;
+    int64_t nrt;  // point tiles
+    int k;
+    int nct;  // centroid tiles
+    int nkc;  // 64-wide k-slices
+    const float4 *cinfo;  // SCREEN: per centroid (||c||^2, h, ||c||, z)
+    const float2 *xinfo;  // SCREEN: per point (||x~||, ||x~ - x||)
+    int32_t *cand;        // SCREEN: [n][TCAND + 1]
+    int32_t *resc_rows;
+    int32_t *fall_rows;
+    int32_t *counters;  // [0] rescore rows, [1] fallback rows, [2] abort flag
+    int32_t *assign;
+    const int32_t *nx;  // SQ8: centred ||x||^2
+    const int32_t *nc;  // SQ8: centred ||c||^2
+    float *dist;        // SQ8 (may be null)
+};
+
+// ------------------------------------------------------------- PTX helpers
+__device__ __forceinline__ uint32_t smem_u32(const void *p) {
+    return (uint32_t)__cvta_generic_to_shared(p);
+}
+__device__ __forceinline__ unsigned long long globaltimer() {
+    unsigned long long t;
+    asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+    return t;
+}
+__device__ __forceinline__ void mbar_init(uint32_t bar, uint32_t count) {
+    asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(bar), "r"(count) : "memory");
+}
+__device__ __forceinline__ void mbar_expect_tx(uint32_t bar, uint32_t bytes) {
+    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"(bytes)
+                 : "memory");
+}
+__device__ __forceinline__ void mbar_arrive(uint32_t bar) {
+    asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(bar) : "memory");
+}
+__device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
+    uint32_t ok;
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+        "selp.u32 %0, 1, 0, p;\n\t}\n"
+        : "=r"(ok)
+        : "r"(bar), "r"(parity)
+        : "memory");
+    return ok != 0;
+}
+// Bounded wait: false when the abort flag is raised or the limit elapses
+// (the flag is then raised so that every role stops).
+__device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, volatile int32_t *abort_flag) {
+    if (mbar_try_wait(bar, parity)) return true;
+    const unsigned long long t0 = globaltimer();
+    for (uint32_t i = 1;; ++i) {
+        if (mbar_try_wait(bar, parity)) return true;
+        if ((i & 255) == 0) {
+            if (*abort_flag) return false;
+            if (globaltimer() - t0 > WAIT_LIMIT_NS) {
+                *abort_flag = 1;
+                return false;
+            }
+        }
+    }
+}
+__device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap *map, int x, int y,
+                                            uint32_t bar) {
+    asm volatile(
+        "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes"
+        " [%0], [%1, {%2, %3}], [%4];" ::"r"(dst),
+        "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(bar)
+        : "memory");
+}
+__device__ __forceinline__ void tc_fence_before() {
+    asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+}
+__device__ __forceinline__ void tc_fence_after() {
+    asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+}
+__device__ __forceinline__ void tc_commit(uint32_t bar) {
+    asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(
+                     bar)
+                 : "memory");
+}
+__device__ __forceinline__ void tc_mma(uint32_t dtmem, uint64_t adesc, uint64_t bdesc, uint32_t idesc,
+                                       uint32_t accumulate) {
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "setp.ne.b32 p, %4, 0;\n\t"
+        "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}\n" ::"r"(dtmem),
+        "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate)
+        : "memory");
+}
+// 32 lanes x 32 consecutive 32-bit columns: thread i receives lane (base + i).
+__device__ __forceinline__ void tmem_ld32(uint32_t taddr, uint32_t (&v)[32]) {
+    asm volatile(
+        "tcgen05.ld.sync.aligned.32x32b.x32.b32 "
+        "{%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15, "
+        "%16, %17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, %29, %30, %31}, [%32];"
+        : "=r"(v[0]), "=r"(v[1]), "=r"(v[2]), "=r"(v[3]), "=r"(v[4]), "=r"(v[5]), "=r"(v[6]),
+          "=r"(v[7]), "=r"(v[8]), "=r"(v[9]), "=r"(v[10]), "=r"(v[11]), "=r"(v[12]), "=r"(v[13]),
+          "=r"(v[14]), "=r"(v[15]), "=r"(v[16]), "=r"(v[17]), "=r"(v[18]), "=r"(v[19]),
+          "=r"(v[20]), "=r"(v[21]), "=r"(v[22]), "=r"(v[23]), "=r"(v[24]), "=r"(v[25]),
+          "=r"(v[26]), "=r"(v[27]), "=r"(v[28]), "=r"(v[29]), "=r"(v[30]), "=r"(v[31])
+        : "r"(taddr)
+        : "memory");
+    asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+}
+
+// Shared-memory matrix descriptor: K-major operand, 128-byte swizzle, rows of
+// 128 bytes in 8-row (1024-byte) groups as written by TMA.  The start address
+// advances by 32 bytes per K=16 step inside the swizzle row.
+__device__ __forceinline__ uint64_t sw128_desc(uint32_t saddr) {
+    uint64_t d = (uint64_t)((saddr & 0x3FFFFu) >> 4);  // start address
+    d |= (uint64_t)1 << 16;                            // leading byte offset (unused here)
+    d |= (uint64_t)(1024 >> 4) << 32;                  // stride byte offset: 8 rows x 128 B
+    d |= (uint64_t)1 << 46;                            // descriptor version (sm_100 family)
+    d |= (uint64_t)2 << 61;                            // 128-byte swizzle
+    return d;
+}
+
+// Instruction descriptor, kind::f16: D fp32, A/B bf16, both K-major,
+// N = 256, M = 128.
+constexpr uint32_t IDESC = (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(BN >> 3) << 17) |
+                           ((uint32_t)(BM >> 4) << 24);
+
+// ------------------------------------------------------ screening row state
+struct ScreenRow {
+    float L[TCAND];
+    int J[TCAND];
+    float umin, lev;
+    float a, r;  // ||x~||, ||x~ - x||
+};
+
+__device__ __forceinline__ void screen_init(ScreenRow &s, float2 xi) {
+#pragma unroll
+    for (int t = 0; t < TCAND; ++t) {
+        s.L[t] = INFINITY;
+        s.J[t] = -1;
+    }
+    s.umin = INFINITY;
+    s.lev = INFINITY;
+    s.a = xi.x;
+    s.r = xi.y;
+}
+
+__device__ __forceinline__ void screen_take(ScreenRow &s, float acc, float4 ci, int j) {
+    const float sv = fmaf(-2.0f, acc, ci.x);        // ||c||^2 - 2 x~.c~
+    float t = fmaf(s.a, ci.y, ci.w);                 // bound / 2
+    t = fmaf(s.r, ci.z, t);
+    const float L = fmaf(-2.0f, t, sv);
+    const float U = fmaf(2.0f, t, sv);
+    s.umin = fminf(s.umin, U);
+    if (L < s.L[TCAND - 1]) {
+        s.lev = fminf(s.lev, s.L[TCAND - 1]);
+        // insertion into the sorted list (strict <: earlier index first on ties)
+        if (L < s.L[2]) {
+            s.L[3] = s.L[2];
+            s.J[3] = s.J[2];
+            if (L < s.L[1]) {
+                s.L[2] = s.L[1];
+                s.J[2] = s.J[1];
+                if (L < s.L[0]) {
+                    s.L[1] = s.L[0];
+                    s.J[1] = s.J[0];
+                    s.L[0] = L;
+                    s.J[0] = j;
+                } else {
+                    s.L[1] = L;
+                    s.J[1] = j;
+                }
+            } else {
+                s.L[2] = L;
+                s.J[2] = j;
+            }
+        } else {
+            s.L[3] = L;
+            s.J[3] = j;
+        }
+    } else {
+        s.lev = fminf(s.lev, L);
+    }
+}
+
+template <int MODE>
+__global__ void __launch_bounds__(THREADS, 1)
+    tc_assign_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
+                     const TcParams p) {
+    extern __shared__ uint8_t smem_raw[];
+    const uint32_t raw = smem_u32(smem_raw);
+    const uint32_t base = (raw + 1023u) & ~1023u;
+    uint8_t *smem = smem_raw + (base - raw);
+    const uint32_t sA = base;
+    const uint32_t sB = base + STAGES * A_STAGE;
+    uint64_t *bars = reinterpret_cast<uint64_t *>(smem + (size_t)STAGES * (A_STAGE + B_STAGE));
+    const uint32_t bar0 = smem_u32(bars);
+    auto full_bar = [&](int s) { return bar0 + 8u * s; };
+    auto empty_bar = [&](int s) { return bar0 + 8u * (STAGES + s); };
+    auto tfull_bar = [&](int b) { return bar0 + 8u * (2 * STAGES + b); };
+    auto tempty_bar = [&](int b) { return bar0 + 8u * (2 * STAGES + 2 + b); };
+    uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(bars + 2 * STAGES + 4);
+
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    volatile int32_t *abort_flag = p.counters + 2;
+
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < STAGES; ++s) {
+            mbar_init(full_bar(s), 1);
+            mbar_init(empty_bar(s), 1);
+        }
+        for (int b = 0; b < 2; ++b) {
+            mbar_init(tfull_bar(b), 1);
+            mbar_init(tempty_bar(b), EPI_WARPS * 32);
+        }
+        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+        asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmA)) : "memory");
+        asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmB)) : "memory");
+    }
+    if (warp == 1) {
+        asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
+                         smem_u32(tmem_slot)),
+                     "r"(512)
+                     : "memory");
+        asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = *tmem_slot;
+
+    if (warp == 0) {
+        if (lane == 0) {  // ---------------------------------------- TMA producer
+            uint32_t it = 0;
+            for (int64_t rt = blockIdx.x; rt < p.nrt; rt += gridDim.x)
+                for (int ct = 0; ct < p.nct; ++ct)
+                    for (int kc = 0; kc < p.nkc; ++kc, ++it) {
+                        const uint32_t s = it % STAGES, ph = (it / STAGES) & 1u;
+                        if (!mbar_wait(empty_bar(s), ph ^ 1u, abort_flag)) goto producer_done;
+                        mbar_expect_tx(full_bar(s), A_STAGE + B_STAGE);
+                        tma_load_2d(sA + s * A_STAGE, &tmA, kc * BK, (int)(rt * BM), full_bar(s));
+                        tma_load_2d(sB + s * B_STAGE, &tmB, kc * BK, ct * BN, full_bar(s));
+                    }
+        producer_done:;
+        }
+    } else if (warp == 1) {
+        if (lane == 0) {  // ---------------------------------------- MMA issuer
+            uint32_t it = 0, job = 0;
+            for (int64_t rt = blockIdx.x; rt < p.nrt; rt += gridDim.x)
+                for (int ct = 0; ct < p.nct; ++ct, ++job) {
+                    const uint32_t b = job & 1u, bph = (job >> 1) & 1u;
+                    if (!mbar_wait(tempty_bar(b), bph ^ 1u, abort_flag)) goto mma_done;
+                    tc_fence_after();
+                    const uint32_t dcol = tmem + b * BN;
+                    for (int kc = 0; kc < p.nkc; ++kc, ++it) {
+                        const uint32_t s = it % STAGES, ph = (it / STAGES) & 1u;
+                        if (!mbar_wait(full_bar(s), ph, abort_flag)) goto mma_done;
+                        tc_fence_after();
+                        const uint64_t ad = sw128_desc(sA + s * A_STAGE);
+                        const uint64_t bd = sw128_desc(sB + s * B_STAGE);
+#pragma unroll
+                        for (int kk = 0; kk < BK / 16; ++kk)
+                            tc_mma(dcol, ad + 2u * kk, bd + 2u * kk, IDESC, (kc | kk) != 0);
+                        tc_commit(empty_bar(s));
+                    }
+                    tc_commit(tfull_bar(b));
+                }
+        mma_done:;
+        }
+    } else {  // ------------------------------------------------------- epilogue
+        const int q = warp & 3;  // TMEM lane quarter this warp may access
+        const int rin = q * 32 + lane;
+        uint32_t job = 0;
+        for (int64_t rt = blockIdx.x; rt < p.nrt; rt += gridDim.x) {
+            const int64_t row = rt * BM + rin;
+            const bool valid = row < p.n;
+            ScreenRow sr;
+            int32_t best = 0x7fffffff, besti = 0;
+            int32_t nxr = 0;
+            if (MODE == MODE_SCREEN)
+                screen_init(sr, valid ? p.xinfo[row] : make_float2(0.f, 0.f));
+            else
+                nxr = valid ? p.nx[row] : 0;
+            for (int ct = 0; ct < p.nct; ++ct, ++job) {
+                const uint32_t b = job & 1u, bph = (job >> 1) & 1u;
+                const bool ok = mbar_wait(tfull_bar(b), bph, abort_flag);
+                if (!__all_sync(0xffffffffu, ok)) goto epi_done;
+                tc_fence_after();
+                const uint32_t taddr = tmem + ((uint32_t)(q * 32) << 16) + b * BN;
+#pragma unroll 1
+                for (int c = 0; c < BN / 32; ++c) {
+                    const int j0 = ct * BN + c * 32;
+                    if (j0 >= p.k) break;  // warp-uniform
+                    uint32_t v[32];
+                    tmem_ld32(taddr + c * 32, v);
+                    if (MODE == MODE_SCREEN) {
+#pragma unroll
+                        for (int i = 0; i < 32; ++i) {
+                            const int j = j0 + i;
+                            if (j < p.k) screen_take(sr, __uint_as_float(v[i]), __ldg(p.cinfo + j), j);
+                        }
+                    } else {
+#pragma unroll
+                        for (int i = 0; i < 32; ++i) {
+                            const int j = j0 + i;
+                            if (j < p.k) {
+                                const int32_t dot = __float2int_rn(__uint_as_float(v[i]));
+                                const int32_t dd = nxr + __ldg(p.nc + j) - 2 * dot;
+                                if (dd < best) {
+                                    best = dd;
+                                    besti = j;
+                                }
+                            }
+                        }
+                    }
+                }
+                tc_fence_before();
+                mbar_arrive(tempty_bar(b));
+            }
+            if (valid) {
+                if (MODE == MODE_SCREEN) {
+                    int ncert = 0;
+#pragma unroll
+                    for (int t = 0; t < TCAND; ++t) ncert += (sr.L[t] <= sr.umin) ? 1 : 0;
+                    const bool overflow = !(sr.lev > sr.umin);
+                    if (!overflow && ncert == 1) {
+                        p.assign[row] = sr.J[0];
+                    } else if (!overflow && ncert >= 2) {
+                        int32_t *cr = p.cand + row * (TCAND + 1);
+#pragma unroll
+                        for (int t = 0; t < TCAND; ++t) cr[t] = sr.J[t];
+                        cr[TCAND] = ncert;
+                        p.assign[row] = sr.J[0];
+                        p.resc_rows[atomicAdd(&p.counters[0], 1)] = (int32_t)row;
+                    } else {
+                        p.assign[row] = sr.J[0] >= 0 ? sr.J[0] : 0;
+                        p.fall_rows[atomicAdd(&p.counters[1], 1)] = (int32_t)row;
+                    }
+                } else {
+                    p.assign[row] = besti;
+                    if (p.dist) p.dist[row] = (float)best;
+                }
+            }
+        }
+    epi_done:;
+    }
+    tc_fence_before();
+    __syncthreads();
+    if (warp == 1) {
+        __syncwarp();
+        tc_fence_after();
+        asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(512)
+                     : "memory");
+    }
+}
+
+// ------------------------------------------------------------- preparation
+// fp32 points -> bf16 screening copy (row stride dp) and per-row
+// (||x~||, ||x~ - x||), both rounded up.  One warp per row.
+__global__ void screen_prep_f32_kernel(const float *__restrict__ X, int64_t n, int d, int dp,
+                                       __nv_bfloat16 *__restrict__ xs, float2 *__restrict__ xinfo) {
+    const int lane = threadIdx.x & 31;
+    const int64_t warp = (blockIdx.x * (int64_t)blockDim.x + threadIdx.x) >> 5;
+    const int64_t nw = ((int64_t)gridDim.x * blockDim.x) >> 5;
+    for (int64_t r = warp; r < n; r += nw) {
+        double a2 = 0.0, r2 = 0.0;
+        for (int i = lane; i < d; i += 32) {
+            const float x = X[r * d + i];
+            const __nv_bfloat16 xb = __float2bfloat16_rn(x);
+            xs[r * dp + i] = xb;
+            const double xf = (double)__bfloat162float(xb);
+            a2 += xf * xf;
+            r2 += (xf - (double)x) * (xf - (double)x);
+        }
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) {
+            a2 += __shfl_xor_sync(0xffffffffu, a2, o);
+            r2 += __shfl_xor_sync(0xffffffffu, r2, o);
+        }
+        if (lane == 0)
+            xinfo[r] = make_float2(__double2float_ru(sqrt(a2) * (1.0 + 1e-6)),
+                                   __double2float_ru(sqrt(r2) * (1.0 + 1e-6)));
+    }
+}
+
+// bf16 points: optional padded copy (when the row stride is not a multiple of
+// 16 bytes) and (||x||, 0): the points are the screening operand exactly.
+__global__ void screen_prep_bf16_kernel(const uint16_t *__restrict__ X, int64_t n, int d, int dp,
+                                        uint16_t *__restrict__ xs, float2 *__restrict__ xinfo) {
+    const int lane = threadIdx.x & 31;
+    const int64_t warp = (blockIdx.x * (int64_t)blockDim.x + threadIdx.x) >> 5;
+    const int64_t nw = ((int64_t)gridDim.x * blockDim.x) >> 5;
+    for (int64_t r = warp; r < n; r += nw) {
+        double a2 = 0.0;
+        for (int i = lane; i < d; i += 32) {
+            const uint16_t v = X[r * d + i];
+            if (xs) xs[r * dp + i] = v;
+            const double xf = (double)__uint_as_float(((uint32_t)v) << 16);
+            a2 += xf * xf;
+        }
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) a2 += __shfl_xor_sync(0xffffffffu, a2, o);
+        if (lane == 0) xinfo[r] = make_float2(__double2float_ru(sqrt(a2) * (1.0 + 1e-6)), 0.0f);
+    }
+}
+
+// SQ8 codes -> centred bf16 (code - 128, exact) and centred ||x||^2 (exact).
+__global__ void screen_prep_sq8_kernel(const uint8_t *__restrict__ X, int64_t n, int d, int dp,
+                                       __nv_bfloat16 *__restrict__ xs, int32_t *__restrict__ nx) {
+    const int lane = threadIdx.x & 31;
+    const int64_t warp = (blockIdx.x * (int64_t)blockDim.x + threadIdx.x) >> 5;
+    const int64_t nw = ((int64_t)gridDim.x * blockDim.x) >> 5;
+    for (int64_t r = warp; r < n; r += nw) {
+        int32_t s = 0;
+        for (int i = lane; i < d; i += 32) {
+            const int32_t v = (int32_t)X[r * d + i] - 128;
+            xs[r * dp + i] = __int2bfloat16_rn(v);
+            s += v * v;
+        }
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
+        if (lane == 0) nx[r] = s;
+    }
+}
+
+// Centroids (fp32) -> bf16 operand + (||c||^2, h, ||c||, z) with
+// h = e + (eps_acc + eps_s) (||c|| + e), e = ||c~ - c||, z = eps_s ||c||^2 / 2,
+// so that |s~ - s| <= 2 (||x~|| h + ||x~ - x|| ||c|| + z) (see the header).
+__global__ void cprep_f32_kernel(const float *__restrict__ C, int k, int d, int dp, float eps_acc,
+                                 float eps_s, __nv_bfloat16 *__restrict__ cs,
+                                 float4 *__restrict__ cinfo) {
+    const int lane = threadIdx.x & 31;
+    const int warp = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+    const int nw = (gridDim.x * blockDim.x) >> 5;
+    for (int j = warp; j < k; j += nw) {
+        double c2 = 0.0, e2 = 0.0;
+        for (int i = lane; i < d; i += 32) {
+            const float c = C[(int64_t)j * d + i];
+            const __nv_bfloat16 cb = __float2bfloat16_rn(c);
+            cs[(int64_t)j * dp + i] = cb;
+            const double cf = (double)__bfloat162float(cb);
+            c2 += (double)c * (double)c;
+            e2 += (cf - (double)c) * (cf - (double)c);
+        }
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) {
+            c2 += __shfl_xor_sync(0xffffffffu, c2, o);
+            e2 += __shfl_xor_sync(0xffffffffu, e2, o);
+        }
+        if (lane == 0) {
+            const double up = 1.0 + 1e-6;
+            const double cn = sqrt(c2), e = sqrt(e2) * up;
+            const double g = (cn + e) * up;
+            const double h = (e + ((double)eps_acc + (double)eps_s) * g) * up;
+            const double z = 0.5 * (double)eps_s * c2 * up;
+            cinfo[j] = make_float4(__double2float_rn(c2), __double2float_ru(h),
+                                   __double2float_ru(cn * up), __double2float_ru(z));
+        }
+    }
+}
+
+__global__ void cprep_sq8_kernel(const uint8_t *__restrict__ C, int k, int d, int dp,
+                                 __nv_bfloat16 *__restrict__ cs, int32_t *__restrict__ nc) {
+    const int lane = threadIdx.x & 31;
+    const int warp = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+    const int nw = (gridDim.x * blockDim.x) >> 5;
+    for (int j = warp; j < k; j += nw) {
+        int32_t s = 0;
+        for (int i = lane; i < d; i += 32) {
+            const int32_t v = (int32_t)C[(int64_t)j * d + i] - 128;
+            cs[(int64_t)j * dp + i] = __int2bfloat16_rn(v);
+            s += v * v;
+        }
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
+        if (lane == 0) nc[j] = s;
+    }
+}
+
+// ------------------------------------------------------------ fp32 rescoring
+template <typename TX>
+__device__ __forceinline__ float ldx(const TX *p);
+template <>
+__device__ __forceinline__ float ldx<float>(const float *p) {
+    return __ldg(p);
+}
+template <>
+__device__ __forceinline__ float ldx<uint16_t>(const uint16_t *p) {
+    return __uint_as_float(((uint32_t)__ldg(p)) << 16);
+}
+
+template <typename TX>
+__device__ __forceinline__ float warp_sqdist(const TX *x, const float *c, int d, int lane) {
+    float s = 0.0f;
+    for (int i = lane; i < d; i += 32) {
+        const float t = __fsub_rn(ldx<TX>(x + i), __ldg(c + i));
+        s = __fmaf_rn(t, t, s);
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
+    return s;
+}
+
+// One warp per listed row: exact fp32 distances to its screen candidates.
+template <typename TX>
+__global__ void rescore_kernel(const TX *__restrict__ X, int d, const float *__restrict__ C,
+                               const int32_t *__restrict__ rows, const int32_t *__restrict__ count,
+                               const int32_t *__restrict__ cand, int32_t *__restrict__ assign) {
+    const int lane = threadIdx.x & 31;
+    const int64_t warp = (blockIdx.x * (int64_t)blockDim.x + threadIdx.x) >> 5;
+    const int64_t nw = ((int64_t)gridDim.x * blockDim.x) >> 5;
+    const int64_t cnt = *count;
+    for (int64_t i = warp; i < cnt; i += nw) {
+        const int64_t r = rows[i];
+        const int32_t *cr = cand + r * (TCAND + 1);
+        const int nc = cr[TCAND];
+        float bd = INFINITY;
+        int bj = 0x7fffffff;
+        for (int t = 0; t < nc; ++t) {
+            const int j = cr[t];
+            const float dd = warp_sqdist<TX>(X + r * d, C + (int64_t)j * d, d, lane);
+            if (dd < bd || (dd == bd && j < bj)) {
+                bd = dd;
+                bj = j;
+            }
+        }
+        if (lane == 0) assign[r] = bj;
+    }
+}
+
+// dist[r] = fp32 sum of squared differences to the assigned centroid.
+template <typename TX>
+__global__ void assigned_dist_kernel(const TX *__restrict__ X, int64_t n, int d,
+                                     const float *__restrict__ C, const int32_t *__restrict__ assign,
+                                     float *__restrict__ dist) {
+    const int lane = threadIdx.x & 31;
+    const int64_t warp = (blockIdx.x * (int64_t)blockDim.x + threadIdx.x) >> 5;
+    const int64_t nw = ((int64_t)gridDim.x * blockDim.x) >> 5;
+    for (int64_t r = warp; r < n; r += nw) {
+        const float dd = warp_sqdist<TX>(X + r * d, C + (int64_t)assign[r] * d, d, lane);
+        if (lane == 0) dist[r] = dd;
+    }
+}
+
+__global__ void add_stats_kernel(const int32_t *__restrict__ counters, int64_t *__restrict__ stats) {
+    stats[0] += counters[0];
+    stats[1] += counters[1];
+    stats[2] |= counters[2];
+}
+
+// ------------------------------------------------------------------ host side
+PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
+    static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+    static std::once_flag once;
+    std::call_once(once, [] {
+        void *p = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault,
+                                             &q) == cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
+    });
+    return fn;
+}
+
+// 2D bf16 map over [rows][cols] (row stride `stride_elems`), box = box_rows x 64.
+int make_map(CUtensorMap *m, const void *ptr, int64_t rows, int cols, int stride_elems,
+             int box_rows) {
+    auto fn = encode_fn();
+    if (!fn) return set_error(SKM_ERR_CUDA, "cuTensorMapEncodeTiled entry point not found");
+    cuuint64_t gdim[2] = {(cuuint64_t)cols, (cuuint64_t)rows};
+    cuuint64_t gstride[1] = {(cuuint64_t)stride_elems * 2};
+    cuuint32_t box[2] = {(cuuint32_t)BK, (cuuint32_t)box_rows};
+    cuuint32_t estr[2] = {1, 1};
+    CUresult r = fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void *>(ptr), gdim, gstride,
+                    box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                    CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    if (r != CUDA_SUCCESS) return set_error(SKM_ERR_CUDA, "cuTensorMapEncodeTiled failed (%d)", (int)r);
+    return SKM_OK;
+}
+
+int device_sms() {
+    int dev = 0, sms = 0;
+    cudaGetDevice(&dev);
+    cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+    return sms > 0 ? sms : 148;
+}
+
+template <int MODE>
+int launch_tc(const void *xs, int64_t n, int dp, int d, const void *cs, int k, const TcParams &p0,
+              cudaStream_t st) {
+    static std::once_flag attr_once[2];
+    static cudaError_t attr_err[2] = {cudaSuccess, cudaSuccess};
+    std::call_once(attr_once[MODE], [] {
+        attr_err[MODE] = cudaFuncSetAttribute(tc_assign_kernel<MODE>,
+                                              cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                              (int)SMEM_BYTES);
+    });
+    if (attr_err[MODE] != cudaSuccess)
+        return set_error(SKM_ERR_CUDA, "cudaFuncSetAttribute: %s", cudaGetErrorString(attr_err[MODE]));
+    CUtensorMap ma, mb;
+    SKM_TRY(make_map(&ma, xs, n, d, dp, BM));
+    SKM_TRY(make_map(&mb, cs, k, d, dp, BN));
+    TcParams p = p0;
+    p.n = n;
+    p.nrt = cdiv(n, BM);
+    p.k = k;
+    p.nct = (int)cdiv(k, BN);
+    p.nkc = (int)cdiv(d, BK);
+    const int grid = (int)std::min<int64_t>(device_sms(), p.nrt);
+    tc_assign_kernel<MODE><<<grid, THREADS, SMEM_BYTES, st>>>(ma, mb, p);
+    SKM_CUDA_TRY(launched());
+    return SKM_OK;
+}
+
+int grid_warps(int64_t items) {
+    int64_t b = (items * 32 + 255) / 256;
+    const int64_t cap = 152LL * 8;
+    return (int)(b < 1 ? 1 : (b > cap ? cap : b));
+}
+
+inline int round8(int d) { return (d + 7) & ~7; }
+
+}  // namespace
+
+// ------------------------------------------------------------- public (internal)
+size_t tc_screen_bytes(int repr, int64_t n, int d, const void *x) {
+    Carver cv(nullptr, 0);
+    const int dp = round8(d);
+    switch (repr) {
+    case SKM_REPR_F32:
+        cv.take<uint16_t>((size_t)n * dp);
+        cv.take<float2>(n);
+        break;
+    case SKM_REPR_SQ8:
+        if (d > TC_SQ8_MAX_D) return 0;
+        cv.take<uint16_t>((size_t)n * dp);
+        cv.take<int32_t>(n);
+        break;
+    case SKM_REPR_BF16:
+        if (d % 8 != 0 || ((uintptr_t)x & 15) != 0) cv.take<uint16_t>((size_t)n * dp);
+        cv.take<float2>(n);
+        break;
+    default:
+        return 0;
+    }
+    return cv.off;
+}
+
+struct ScreenView {
+    const void *xs = nullptr;
+    const float2 *xinfo = nullptr;
+    const int32_t *nx = nullptr;
+};
+
+static ScreenView screen_view(int repr, int64_t n, int d, const void *x, const void *screen) {
+    ScreenView v;
+    Carver cv(const_cast<void *>(screen), SIZE_MAX);
+    const int dp = round8(d);
+    switch (repr) {
+    case SKM_REPR_F32:
+        v.xs = cv.take<uint16_t>((size_t)n * dp);
+        v.xinfo = cv.take<float2>(n);
+        break;
+    case SKM_REPR_SQ8:
+        v.xs = cv.take<uint16_t>((size_t)n * dp);
+        v.nx = cv.take<int32_t>(n);
+        break;
+    case SKM_REPR_BF16:
+        if (d % 8 != 0 || ((uintptr_t)x & 15) != 0)
+            v.xs = cv.take<uint16_t>((size_t)n * dp);
+        else
+            v.xs = x;
+        v.xinfo = cv.take<float2>(n);
+        break;
+    }
+    return v;
+}
+
+int tc_screen_prep(const skm_data *x, void *screen, cudaStream_t st) {
+    const int64_t n = x->n;
+    const int d = x->d, dp = round8(d);
+    ScreenView v = screen_view(x->repr, n, d, x->x, screen);
+    const int g = grid_warps(n);
+    switch (x->repr) {
+    case SKM_REPR_F32:
+        screen_prep_f32_kernel<<<g, 256, 0, st>>>(static_cast<const float *>(x->x), n, d, dp,
+                                                  (__nv_bfloat16 *)v.xs, (float2 *)v.xinfo);
+        break;
+    case SKM_REPR_SQ8:
+        screen_prep_sq8_kernel<<<g, 256, 0, st>>>(static_cast<const uint8_t *>(x->x), n, d, dp,
+                                                  (__nv_bfloat16 *)v.xs, (int32_t *)v.nx);
+        break;
+    case SKM_REPR_BF16:
+        screen_prep_bf16_kernel<<<g, 256, 0, st>>>(static_cast<const uint16_t *>(x->x), n, d, dp,
+                                                   v.xs == x->x ? nullptr : (uint16_t *)v.xs,
+                                                   (float2 *)v.xinfo);
+        break;
+    default:
+        return set_error(SKM_ERR_INVALID_ARG, "no screening copy for repr %d", x->repr);
+    }
+    SKM_CUDA_TRY(launched());
+    return SKM_OK;
+}
+
+void tc_plan(int repr, int64_t n, int d, int k, const void *x, const void *screen, Carver &cv,
+             TcAssignBufs &b) {
+    b.stats = cv.take<int64_t>(4);
+    b.counters = cv.take<int32_t>(4);
+    const int dp = round8(d);
+    const bool dense = repr == SKM_REPR_F32 || repr == SKM_REPR_BF16 ||
+                       (repr == SKM_REPR_SQ8 && d <= TC_SQ8_MAX_D);
+    if (!dense) return;
+    if (!screen) {
+        const size_t sb = tc_screen_bytes(repr, n, d, x);
+        b.screen = cv.take<uint8_t>(sb);
+    }
+    b.cs = cv.take<uint16_t>((size_t)k * dp);
+    if (repr == SKM_REPR_SQ8) {
+        b.nc = cv.take<int32_t>(k);
+    } else {
+        b.cinfo = cv.take<float4>(k);
+        b.cand = cv.take<int32_t>((size_t)n * (TCAND + 1));
+        b.resc_rows = cv.take<int32_t>(n);
+        b.fall_rows = cv.take<int32_t>(n);
+    }
+}
+
+int tc_init_stats(TcAssignBufs &b, cudaStream_t st) {
+    SKM_CUDA_TRY(cudaMemsetAsync(b.stats, 0, sizeof(int64_t) * 4, st));
+    return SKM_OK;
 }
 
 int tc_assign_float(const skm_data *x, const float *C, int k, int32_t *assign, float *dist,
                     TcAssignBufs &b, cudaStream_t st) {
-    (void)b;
-    if (x->repr == SKM_REPR_BF16)
-        SKM_CUDA_TRY(launch_assign_exact_bf16(static_cast<const uint16_t *>(x->x), x->n, x->d, C, k,
-                                              assign, dist, st));
-    else
-        SKM_CUDA_TRY(launch_assign_exact_f32(static_cast<const float *>(x->x), x->n, x->d, C, k,
-                                             assign, dist, st));
+    const int64_t n = x->n;
+    const int d = x->d, dp = round8(d);
+    const bool bf16 = x->repr == SKM_REPR_BF16;
+    const void *screen = x->screen;
+    if (!screen) {
+        skm_data tmp = *x;
+        SKM_TRY(tc_screen_prep(&tmp, b.screen, st));
+        screen = b.screen;
+    }
+    ScreenView v = screen_view(x->repr, n, d, x->x, screen);
+    const int nkc = (int)cdiv(d, BK);
+    const float eps_acc = (float)((nkc * (BK / 16) + 4) * 0x1p-18);
+    const float eps_s = 0x1p-21f;
+    cprep_f32_kernel<<<grid_warps(k), 256, 0, st>>>(C, k, d, dp, eps_acc, eps_s,
+                                                    (__nv_bfloat16 *)b.cs, b.cinfo);
+    SKM_CUDA_TRY(launched());
+    SKM_CUDA_TRY(cudaMemsetAsync(b.counters, 0, sizeof(int32_t) * 4, st));
+    TcParams p{};
+    p.cinfo = b.cinfo;
+    p.xinfo = v.xinfo;
+    p.cand = b.cand;
+    p.resc_rows = b.resc_rows;
+    p.fall_rows = b.fall_rows;
+    p.counters = b.counters;
+    p.assign = assign;
+    SKM_TRY(launch_tc<MODE_SCREEN>(v.xs, n, dp, d, b.cs, k, p, st));
+    const int gw = grid_warps(n);
+    if (bf16) {
+        const uint16_t *X = static_cast<const uint16_t *>(x->x);
+        rescore_kernel<uint16_t><<<gw, 256, 0, st>>>(X, d, C, b.resc_rows, b.counters, b.cand, assign);
+        SKM_CUDA_TRY(launched());
+        SKM_CUDA_TRY(launch_assign_exact_rows(X, 1, b.fall_rows, b.counters + 1, n, d, C, k, assign,
+                                              nullptr, st));
+        if (dist) {
+            assigned_dist_kernel<uint16_t><<<gw, 256, 0, st>>>(X, n, d, C, assign, dist);
+            SKM_CUDA_TRY(launched());
+        }
+    } else {
+        const float *X = static_cast<const float *>(x->x);
+        rescore_kernel<float><<<gw, 256, 0, st>>>(X, d, C, b.resc_rows, b.counters, b.cand, assign);
+        SKM_CUDA_TRY(launched());
+        SKM_CUDA_TRY(launch_assign_exact_rows(X, 0, b.fall_rows, b.counters + 1, n, d, C, k, assign,
+                                              nullptr, st));
+        if (dist) {
+            assigned_dist_kernel<float><<<gw, 256, 0, st>>>(X, n, d, C, assign, dist);
+            SKM_CUDA_TRY(launched());
+        }
+    }
+    add_stats_kernel<<<1, 1, 0, st>>>(b.counters, b.stats);
+    SKM_CUDA_TRY(launched());
     return SKM_OK;
 }
 
-int tc_assign_sq8(const skm_data *x, const uint8_t *C, int k, const int32_t *nx,
-                  const int32_t *nc, int32_t *assign, float *dist, TcAssignBufs &b,
+int tc_assign_sq8(const skm_data *x, const uint8_t *C, int k, int32_t *nx_plain,
+                  int32_t *nc_plain, int32_t *assign, float *dist, TcAssignBufs &b,
                   cudaStream_t st) {
-    (void)b;
-    SKM_CUDA_TRY(launch_assign_sq8_simt(static_cast<const uint8_t *>(x->x), x->n, x->d, C, k, nx,
-                                        nc, assign, dist, st));
+    const int64_t n = x->n;
+    const int d = x->d, dp = round8(d);
+    if (d > TC_SQ8_MAX_D) {  // the bf16 accumulation is exact only up to d = 1024
+        const uint8_t *X = static_cast<const uint8_t *>(x->x);
+        SKM_CUDA_TRY(launch_row_sqnorm_u8(X, n, d, nx_plain, st));
+        SKM_CUDA_TRY(launch_row_sqnorm_u8(C, k, d, nc_plain, st));
+        SKM_CUDA_TRY(launch_assign_sq8_simt(X, n, d, C, k, nx_plain, nc_plain, assign, dist, st));
+        return SKM_OK;
+    }
+    const void *screen = x->screen;
+    if (!screen) {
+        skm_data tmp = *x;
+        SKM_TRY(tc_screen_prep(&tmp, b.screen, st));
+        screen = b.screen;
+    }
+    ScreenView v = screen_view(x->repr, n, d, x->x, screen);
+    cprep_sq8_kernel<<<grid_warps(k), 256, 0, st>>>(C, k, d, dp, (__nv_bfloat16 *)b.cs, b.nc);
+    SKM_CUDA_TRY(launched());
+    SKM_CUDA_TRY(cudaMemsetAsync(b.counters, 0, sizeof(int32_t) * 4, st));
+    TcParams p{};
+    p.counters = b.counters;
+    p.assign = assign;
+    p.nx = v.nx;
+    p.nc = b.nc;
+    p.dist = dist;
+    SKM_TRY(launch_tc<MODE_SQ8>(v.xs, n, dp, d, b.cs, k, p, st));
+    add_stats_kernel<<<1, 1, 0, st>>>(b.counters, b.stats);
+    SKM_CUDA_TRY(launched());
     return SKM_OK;
 }
 
-void tc_read_stats(const TcAssignBufs &b, skm_stats *st_host, cudaStream_t st) {
-    (void)b; (void)st; (void)st_host;
+int tc_read_stats(const TcAssignBufs &b, skm_stats *st_host, cudaStream_t st) {
+    int64_t h[4] = {0, 0, 0, 0};
+    SKM_CUDA_TRY(cudaMemcpyAsync(h, b.stats, sizeof(h), cudaMemcpyDeviceToHost, st));
+    SKM_CUDA_TRY(cudaStreamSynchronize(st));
+    if (st_host) {
+        st_host->rescored_rows = h[0];
+        st_host->fallback_rows = h[1];
+    }
+    if (h[2]) return set_error(SKM_ERR_TIMEOUT, "a tensor-core pipeline wait exceeded its limit");
+    return SKM_OK;
 }
 
 }  // namespace skm

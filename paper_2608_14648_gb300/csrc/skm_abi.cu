@@ -59,21 +59,21 @@ static int check_data(const skm_data *x, bool need_codes = true) {
     return SKM_OK;
 }
 
-static int check_k(const skm_data *x, int k) {
+static int check_k(const skm_data *x, int k, bool k_le_n = false) {
     if (k < 1 || k > MAX_K)
         return set_error(k < 1 ? SKM_ERR_INVALID_ARG : SKM_ERR_UNSUPPORTED,
                          "k = %d outside [1, %d]", k, MAX_K);
-    if ((int64_t)k > x->n)
+    if (k_le_n && (int64_t)k > x->n)
         return set_error(SKM_ERR_INVALID_ARG, "k = %d exceeds n = %lld", k, (long long)x->n);
     return SKM_OK;
 }
 
 // ------------------------------------------------------------ workspace plans
 struct AssignBufs {
-    int32_t *nx = nullptr, *nc = nullptr;  // SQ8
+    int32_t *nx = nullptr, *nc = nullptr;  // SQ8 with d > 1024 (__dp4a path)
     uint4 *planes = nullptr;                // RBQ1
     Rbq1CInfo *info = nullptr;
-    TcAssignBufs tc;                        // F32 / BF16 / SQ8 tensor-core screen
+    TcAssignBufs tc;                        // F32 / BF16 / SQ8 tensor-core path
 };
 
 static void plan_assign(const skm_data *x, int k, Carver &cv, AssignBufs &b) {
@@ -81,8 +81,10 @@ static void plan_assign(const skm_data *x, int k, Carver &cv, AssignBufs &b) {
     const int d = x->d;
     switch (x->repr) {
     case SKM_REPR_SQ8:
-        b.nx = cv.take<int32_t>(n);
-        b.nc = cv.take<int32_t>(k);
+        if (d > TC_SQ8_MAX_D) {
+            b.nx = cv.take<int32_t>(n);
+            b.nc = cv.take<int32_t>(k);
+        }
         break;
     case SKM_REPR_RBQ1:
         b.planes = cv.take<uint4>((size_t)k * words_of(d));
@@ -91,7 +93,7 @@ static void plan_assign(const skm_data *x, int k, Carver &cv, AssignBufs &b) {
     default:
         break;
     }
-    tc_plan(x->repr, n, d, k, cv, b.tc);
+    tc_plan(x->repr, n, d, k, x->x, x->screen, cv, b.tc);
 }
 
 struct UpdateBufs {
@@ -107,6 +109,7 @@ static void plan_update(const skm_data *x, int k, Carver &cv, UpdateBufs &b) {
 }
 
 struct FitBufs {
+    uint8_t *screen = nullptr;  // built once per fit when the caller gave none
     AssignBufs a;
     UpdateBufs u;
     float *dist = nullptr;
@@ -118,7 +121,15 @@ struct FitBufs {
 };
 
 static void plan_fit(const skm_data *x, int k, Carver &cv, FitBufs &b) {
-    plan_assign(x, k, cv, b.a);
+    skm_data xs = *x;
+    if (!x->screen) {
+        const size_t sb = tc_screen_bytes(x->repr, x->n, x->d, x->x);
+        if (sb) {
+            b.screen = cv.take<uint8_t>(sb);
+            xs.screen = b.screen ? b.screen : reinterpret_cast<const void *>(1);  // measured
+        }
+    }
+    plan_assign(&xs, k, cv, b.a);
     plan_update(x, k, cv, b.u);
     b.dist = cv.take<float>(x->n);
     b.partials = cv.take<double>(RED_BLOCKS);
@@ -152,14 +163,10 @@ static int do_assign(const skm_data *x, const void *C, int k, const int32_t *pre
         SKM_TRY(tc_assign_float(x, static_cast<const float *>(C), k, assign, dist, b.tc, st));
         (void)prev;
         break;
-    case SKM_REPR_SQ8: {
-        const uint8_t *X = static_cast<const uint8_t *>(x->x);
-        const uint8_t *Cc = static_cast<const uint8_t *>(C);
-        SKM_CUDA_TRY(launch_row_sqnorm_u8(X, n, d, b.nx, st));
-        SKM_CUDA_TRY(launch_row_sqnorm_u8(Cc, k, d, b.nc, st));
-        SKM_TRY(tc_assign_sq8(x, Cc, k, b.nx, b.nc, assign, dist, b.tc, st));
+    case SKM_REPR_SQ8:
+        SKM_TRY(tc_assign_sq8(x, static_cast<const uint8_t *>(C), k, b.nx, b.nc, assign, dist,
+                              b.tc, st));
         break;
-    }
     case SKM_REPR_RBQ1:
         SKM_CUDA_TRY(
             launch_rbq1_cprep(static_cast<const float *>(C), k, d, x->m, b.planes, b.info, st));
@@ -231,7 +238,7 @@ size_t skm_workspace_size(int op, const skm_data *x, int k) {
         break;
     }
     case 2: {
-        if (check_data(x, false) || check_k(x, k)) return 0;
+        if (check_data(x, false) || check_k(x, k, true)) return 0;
         FitBufs b;
         plan_fit(x, k, cv, b);
         break;
@@ -386,6 +393,22 @@ int skm_rbq1_exponent(const float *F, int64_t n, int *e_host, void *ws, size_t w
     return SKM_OK;
 }
 
+size_t skm_screen_bytes(const skm_data *x) {
+    if (check_data(x, false)) return 0;
+    return tc_screen_bytes(x->repr, x->n, x->d, x->x);
+}
+
+int skm_screen_prep(const skm_data *x, void *screen, size_t screen_bytes, void *stream) {
+    SKM_TRY(check_data(x));
+    const size_t need = tc_screen_bytes(x->repr, x->n, x->d, x->x);
+    if (need == 0) return set_error(SKM_ERR_INVALID_ARG, "this representation has no screening copy");
+    if (!screen || screen_bytes < need)
+        return set_error(SKM_ERR_NO_MEMORY, "screen buffer needs %zu bytes", need);
+    if (((uintptr_t)screen & 255) != 0)
+        return set_error(SKM_ERR_INVALID_ARG, "screen buffer must be 256-byte aligned");
+    return tc_screen_prep(x, screen, S(stream));
+}
+
 int skm_assign(const skm_data *x, const void *C, int k, const int32_t *prev_assign,
                int32_t *assign, float *dist, void *ws, size_t ws_bytes, void *stream) {
     SKM_TRY(check_data(x));
@@ -450,7 +473,7 @@ int skm_fit(const skm_fit_config *cfg, const skm_data *x, const void *C_init,
     if (!cfg) return set_error(SKM_ERR_INVALID_ARG, "cfg is NULL");
     SKM_TRY(check_data(x));
     const int k = cfg->k;
-    SKM_TRY(check_k(x, k));
+    SKM_TRY(check_k(x, k, true));
     if (cfg->iters < 0 || cfg->iters > 100000)
         return set_error(SKM_ERR_INVALID_ARG, "iters = %d", cfg->iters);
     if (!C_out || !assign_out) return set_error(SKM_ERR_INVALID_ARG, "C_out and assign_out required");
@@ -465,6 +488,11 @@ int skm_fit(const skm_fit_config *cfg, const skm_data *x, const void *C_init,
     const int d = x->d;
 
     skm_data xd = *x;
+    if (!x->screen && b.screen) {
+        SKM_TRY(tc_screen_prep(x, b.screen, st));
+        xd.screen = b.screen;
+    }
+    SKM_TRY(tc_init_stats(b.a.tc, st));
     int e = 0;
     if (x->repr == SKM_REPR_RBQ1) {
         SKM_CUDA_TRY(launch_rbq1_exponent(x->F, n, b.maxbits, b.e_dev, st));
@@ -511,9 +539,11 @@ int skm_fit(const skm_fit_config *cfg, const skm_data *x, const void *C_init,
         SKM_TRY(do_update(&xd, assign, k, C_out, b.counts, nullptr, e, b.u, st));
     }
     SKM_CUDA_TRY(cudaStreamSynchronize(st));
+    skm_stats local;
+    memset(&local, 0, sizeof(local));
+    SKM_TRY(tc_read_stats(b.a.tc, &local, st));
     if (stats_host) {
-        memset(stats_host, 0, sizeof(*stats_host));
-        tc_read_stats(b.a.tc, stats_host, st);
+        *stats_host = local;
         std::vector<int64_t> cnt(k);
         if (cfg->iters > 0) {
             SKM_CUDA_TRY(cudaMemcpy(cnt.data(), b.counts, sizeof(int64_t) * k,

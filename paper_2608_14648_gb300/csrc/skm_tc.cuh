@@ -1,20 +1,39 @@
-// Assignment for the dense representations (F32, BF16, SQ8): buffers and
-// entry points used by skm_abi.cu.
+// Tensor-core assignment for the dense representations (F32, BF16, SQ8):
+// buffers and entry points used by skm_abi.cu (implemented in k_tc.cu).
 #pragma once
 #include "skm_internal.cuh"
 
 namespace skm {
 
+// Above this d the fp32 accumulator of the bf16-encoded SQ8 dot product can
+// exceed 2^24 and stop being exact; SQ8 then uses the __dp4a kernel.
+constexpr int TC_SQ8_MAX_D = 1024;
+
 struct TcAssignBufs {
-    int64_t *stats = nullptr;  // [0] rescored rows, [1] fallback rows (cumulative)
+    int64_t *stats = nullptr;     // [0] rescored rows, [1] fallback rows, [2] timeout (cumulative)
+    int32_t *counters = nullptr;  // per call: [0] rescore list, [1] fallback list, [2] abort flag
+    uint8_t *screen = nullptr;    // screening copy built per call when the caller gave none
+    uint16_t *cs = nullptr;       // centroid operand, bf16 [k][round8(d)]
+    float4 *cinfo = nullptr;      // F32/BF16: per-centroid bound terms
+    int32_t *nc = nullptr;        // SQ8: centred ||c||^2
+    int32_t *cand = nullptr;      // F32/BF16: [n][5] screen candidates + count
+    int32_t *resc_rows = nullptr;
+    int32_t *fall_rows = nullptr;
 };
 
-void tc_plan(int repr, int64_t n, int d, int k, Carver &cv, TcAssignBufs &b);
+size_t tc_screen_bytes(int repr, int64_t n, int d, const void *x);
+int tc_screen_prep(const skm_data *x, void *screen, cudaStream_t st);
+void tc_plan(int repr, int64_t n, int d, int k, const void *x, const void *screen, Carver &cv,
+             TcAssignBufs &b);
+int tc_init_stats(TcAssignBufs &b, cudaStream_t st);
 int tc_assign_float(const skm_data *x, const float *C, int k, int32_t *assign, float *dist,
                     TcAssignBufs &b, cudaStream_t st);
-int tc_assign_sq8(const skm_data *x, const uint8_t *C, int k, const int32_t *nx,
-                  const int32_t *nc, int32_t *assign, float *dist, TcAssignBufs &b,
+// nx_plain / nc_plain: buffers for the __dp4a path (d > TC_SQ8_MAX_D), filled here.
+int tc_assign_sq8(const skm_data *x, const uint8_t *C, int k, int32_t *nx_plain,
+                  int32_t *nc_plain, int32_t *assign, float *dist, TcAssignBufs &b,
                   cudaStream_t st);
-void tc_read_stats(const TcAssignBufs &b, skm_stats *st_host, cudaStream_t st);
+// Copies the cumulative statistics; returns SKM_ERR_TIMEOUT if a pipeline
+// wait gave up.  Synchronises the stream.
+int tc_read_stats(const TcAssignBufs &b, skm_stats *st_host, cudaStream_t st);
 
 }  // namespace skm

@@ -45,8 +45,9 @@ FAKE = ctypes.c_void_p(0x1000)
 def test_invalid_arguments_are_rejected_before_launch(skm):
     L = skm.lib()
     x = _data(skm)
-    # k > n
-    rc = L.skm_assign(ctypes.byref(x), FAKE, 101, None, FAKE, None, FAKE, 1 << 20, None)
+    # k > n: allowed for a plain assignment, rejected by fit (Forgy needs k points)
+    cfg = skm.FitConfig(101, 3)
+    rc = L.skm_fit(ctypes.byref(cfg), ctypes.byref(x), None, FAKE, FAKE, FAKE, None, None, None, FAKE, 1 << 30, None)
     assert rc == 1 and b"exceeds" in L.skm_last_error()
     # k = 0
     assert L.skm_assign(ctypes.byref(x), FAKE, 0, None, FAKE, None, FAKE, 1 << 20, None) == 1

@@ -60,6 +60,9 @@ def test_assign_f32_vs_oracle(skm, n, d, k):
     a, dist = skm.skm_assign(pts, C.to(DEV))
     a_or, best, second = oracle.assign_f32(X.numpy(), C.numpy())
     _check_f32(a.cpu().numpy(), dist.cpu().numpy(), best, second, a_or, f"f32 n={n} d={d} k={k}")
+    # the same through a screening copy built once
+    a2, dist2 = skm.skm_assign(pts.with_screen(), C.to(DEV))
+    assert torch.equal(a2, a) and torch.equal(dist2, dist)
 
 
 def test_assign_f32_edge_cases(skm):
@@ -101,6 +104,8 @@ def test_fit_f32_tiny_workload(skm):
     idx = synth.forgy_indices(spec.n, spec.k, seed=0)
     pts = skm.Points(skm.REPR_F32, X.to(DEV), spec.d)
     C, a, dist, obj, stats = skm.skm_fit(pts, spec.k, spec.iters, init_idx=idx.to(DEV))
+    print("tiny fit stats", stats)
+    assert stats["fallback_rows"] < 0.01 * spec.n * (spec.iters + 1)
     Co, ao, objo = oracle.lloyd_f32(X.numpy(), X.numpy()[idx.numpy()], spec.iters)
     agree = (a.cpu().numpy() == ao).mean()
     assert agree >= AGREE
@@ -126,7 +131,8 @@ def test_quantize_sq8_bitexact(skm, n, d):
     np.testing.assert_array_equal(Y.cpu().numpy(), oracle.sq8_decode(q["codes"].cpu().numpy(), b, s))
 
 
-@pytest.mark.parametrize("n,d,k", [(2000, 64, 50), (777, 33, 7), (1024, 1024, 129), (300, 5, 300)])
+@pytest.mark.parametrize("n,d,k", [(2000, 64, 50), (777, 33, 7), (1024, 1024, 129), (300, 5, 300),
+                                   (600, 1500, 40), (1000, 1024, 1)])
 def test_assign_update_sq8_bitexact(skm, n, d, k):
     g = np.random.default_rng(n + d)
     Xc = g.integers(0, 256, size=(n, d)).astype(np.uint8)
