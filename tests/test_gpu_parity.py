@@ -233,9 +233,11 @@ def test_project_vs_oracle(skm, n, d, dout):
     Yb = skm.skm_project(X.to(DEV), P.to(DEV), mu.to(DEV), out_dtype=skm.DTYPE_BF16)
     yb = Yb.view(torch.int16).cpu().numpy().view(np.uint16)
     ybo = oracle.round_bf16(Yo)
-    # bf16 of the fp32 result vs bf16 of the fp64 result: equal or 1 ulp apart
-    diff = np.abs(yb.astype(np.int32) - ybo.astype(np.int32))
-    assert diff.max() <= 1 and (diff == 0).mean() > 0.99
+    # bf16 of the fp32 result vs the fp64 result: within half a bf16 ulp of
+    # the value plus the fp32 accumulation error; identical codes for almost all
+    err = np.abs(oracle.bf16_to_f32(yb).astype(np.float64) - Yo)
+    assert np.all(err <= 2.0 ** -8 * np.abs(Yo) + 2e-6 * scale)
+    assert (yb == ybo).mean() > 0.99
 
 
 @pytest.mark.parametrize("n,d,k", [(2000, 256, 100), (777, 64, 13), (300, 32, 300)])
