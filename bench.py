@@ -393,6 +393,47 @@ def run_reference(args):
     print(json.dumps(line), flush=True)
 
 
+def run_case(args):
+    """Small single-operation runs for profiler captures (ncu): `reps` calls
+    of one entry point on a synthetic workload of the given size."""
+    import torch
+
+    import paper_2608_14648_gb300 as skm
+    import synth
+
+    torch.cuda.set_device(0)
+    n, d, k = args.n, args.d, args.k
+    X = synth.gmm_points(n, d, max(2 * k, 16), seed=0, device="cuda")
+    C = X[synth.forgy_indices(n, k, seed=0).cuda()].clone()
+    if args.case in ("assign_f32", "update_f32"):
+        pts = skm.Points(skm.REPR_F32, X, d).with_screen()
+    elif args.case in ("assign_rbq1", "update_rbq1"):
+        pts = skm.rbq1_points(skm.skm_quantize(skm.REPR_RBQ1, X), d)
+    elif args.case in ("assign_sq8", "update_sq8"):
+        q = skm.skm_quantize(skm.REPR_SQ8, X)
+        pts = skm.Points(skm.REPR_SQ8, q["codes"], d).with_screen()
+        C = q["codes"][:k].clone()
+    else:
+        raise SystemExit(f"unknown case {args.case}")
+    wsA = skm.workspace(skm.OP_ASSIGN, pts, k)
+    wsU = skm.workspace(skm.OP_UPDATE, pts, k)
+    a = torch.empty(n, dtype=torch.int32, device="cuda")
+    cnt = torch.zeros(k, dtype=torch.int64, device="cuda")
+    skm.skm_assign(pts, C, k, want_dist=False, ws=wsA, out=a)
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record()
+    for _ in range(args.reps):
+        if args.case.startswith("assign"):
+            skm.skm_assign(pts, C, k, want_dist=False, ws=wsA, out=a)
+        else:
+            skm.skm_update(pts, a, C.clone(), counts=cnt, ws=wsU)
+    e1.record()
+    torch.cuda.synchronize()
+    print(json.dumps({"case": args.case, "n": n, "d": d, "k": k, "reps": args.reps,
+                      "ms_per_call": e0.elapsed_time(e1) / args.reps}))
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -401,7 +442,17 @@ def main():
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--case", default=None,
+                    help="single-operation run for profiling: assign_f32|assign_rbq1|assign_sq8|update_f32|"
+                         "update_rbq1|update_sq8")
+    ap.add_argument("--n", type=int, default=200_000)
+    ap.add_argument("--d", type=int, default=768)
+    ap.add_argument("--k", type=int, default=1000)
+    ap.add_argument("--reps", type=int, default=3)
     args = ap.parse_args()
+    if args.case:
+        run_case(args)
+        return
     if args.warmup < 3:
         print("warning: fewer than 3 warm-up steps", file=sys.stderr)
     if args.impl == "reference":
