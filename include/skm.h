@@ -203,6 +203,27 @@ int skm_screen_prep(const skm_data *x, void *screen, size_t screen_bytes, void *
 int skm_assign(const skm_data *x, const void *C, int k, const int32_t *prev_assign,
                int32_t *assign, float *dist, void *ws, size_t ws_bytes, void *stream);
 
+/* RBQ1 assignment that allocates nothing.  The paper has no counterpart:
+ * this entry point exists for callers that cannot allocate device memory
+ * (code inside a host engine that owns all device memory through its own pool
+ * or budget, or a latency-critical path where cudaMalloc/cudaFree and their
+ * possible device-wide synchronisation are not acceptable).  Same inputs,
+ * outputs and results as skm_assign with x->repr == SKM_REPR_RBQ1; the
+ * per-centroid scratch (SQ4 bit planes and estimator terms) lives in one
+ * file-scope device array of 2.25 MiB that every GPU which loads the
+ * library keeps until exit.
+ *   Limits: k <= 16384 and k * ceil(d/32) <= 131072, else SKM_ERR_UNSUPPORTED
+ *   (nothing is launched).
+ *   The first call on a device looks up the array's device address with that
+ *   device current (cudaGetSymbolAddress) and caches it; make that first call
+ *   before any stream capture.
+ *   All calls share the array and it keeps the last call's contents: calls
+ *   whose work overlaps on the GPU (other streams, other threads) race; order
+ *   them on one stream or synchronise between them.
+ *   No cudaMalloc, cudaFree or allocating library call is made. */
+int skm_assign_rbq1_noalloc(const skm_data *x, const float *C, int k, int32_t *assign, float *dist,
+                            void *stream);
+
 /* ------------------------------------------------------------------------
  * Update, Section 2.3 STEP 3 (and the quantized-domain variants of 3.1).
  *  C_inout (device), per repr as in skm_assign; clusters with no member keep

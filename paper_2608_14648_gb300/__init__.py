@@ -32,7 +32,8 @@ _lib = None
 EXPORTED_SYMBOLS = [
     "skm_last_error", "skm_version", "skm_kernel_launches", "skm_workspace_size", "skm_screen_bytes",
     "skm_screen_prep", "skm_project", "skm_make_rotation",
-    "skm_pca_fit", "skm_quantize", "skm_rbq1_exponent", "skm_assign", "skm_update",
+    "skm_pca_fit", "skm_quantize", "skm_rbq1_exponent", "skm_assign", "skm_assign_rbq1_noalloc",
+    "skm_update",
     "skm_merge_partials", "skm_update_finalize", "skm_fit", "skm_objective", "skm_sq8_decode",
 ]
 
@@ -96,6 +97,7 @@ def lib():
             "skm_quantize": ([i32, vp, i64, i32, vp, vp, vp, sz, vp], i32),
             "skm_rbq1_exponent": ([vp, i64, vp, vp, sz, vp], i32),
             "skm_assign": ([vp, vp, i32, vp, vp, vp, vp, sz, vp], i32),
+            "skm_assign_rbq1_noalloc": ([vp, vp, i32, vp, vp, vp], i32),
             "skm_update": ([vp, vp, i32, vp, vp, vp, vp, sz, vp], i32),
             "skm_merge_partials": ([vp, vp, i64, i32, vp], i32),
             "skm_update_finalize": ([vp, vp, vp, i32, vp, vp], i32),
@@ -263,6 +265,15 @@ def skm_assign(pts: Points, C, k=None, prev_assign=None, want_dist=True, ws=None
     _check(lib().skm_assign(ctypes.byref(pts.ref), _ptr(C), int(k), _ptr(prev_assign), _ptr(assign), _ptr(dist),
                             _ptr(ws), ws.numel(), _stream(stream)))
     return assign, dist
+
+
+def skm_assign_rbq1_noalloc(pts: Points, C, out, dist_out=None, stream=None):
+    """RBQ1 assignment that allocates nothing in the library (fixed device
+    scratch); `out` (int32[n]) and `dist_out` (float[n] or None) are caller
+    tensors."""
+    _check(lib().skm_assign_rbq1_noalloc(ctypes.byref(pts.ref), _ptr(C), C.shape[0], _ptr(out), _ptr(dist_out),
+                                         _stream(stream)))
+    return out, dist_out
 
 
 def skm_update(pts: Points, assign, C_inout, counts=None, partial=None, ws=None, stream=None):
