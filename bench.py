@@ -168,7 +168,7 @@ def run_ours(args):
         et = torch.tensor([e], device=dev)
         dist.all_reduce(et, op=dist.ReduceOp.MIN)
         e = int(et.item())
-    ptsR = skm.rbq1_points(q, DIM, e)
+    ptsR = skm.rbq1_points(q, DIM, e).with_screen()  # e4m3 expansion of the bits, built once
     Cr, _, _, _, _ = skm.skm_fit(ptsR, K, 0, init_idx=idx, want_objective=False, want_dist=False)
     if world > 1:
         dist.broadcast(Cr, 0)
@@ -235,32 +235,50 @@ def run_ours(args):
     ms_step = ms / args.steps
     value = world * 2.0 * N_POINTS * K * args.steps / (ms / 1e3)
 
+    # ---- the AND+popcount 1-bit kernel, timed beside the tensor-core one --------
+    t_pop = None
+    if not args.no_popcount:
+        torch.cuda.synchronize()
+        p0, p1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a_pop = torch.empty_like(aR)
+        skm.skm_assign_rbq1_noalloc(ptsR, Cr, a_pop)
+        p0.record(stream)
+        skm.skm_assign_rbq1_noalloc(ptsR, Cr, a_pop)
+        p1.record(stream)
+        torch.cuda.synchronize()
+        t_pop = p0.elapsed_time(p1)
+
     # ---- roofline of the dominant kernel --------------------------------------
     t_a32 = statistics.mean(a.elapsed_time(b) for a, b in ev["a32"])
     t_aR = statistics.mean(a.elapsed_time(b) for a, b in ev["aR"])
     long_region = ms > 1000.0
     bf16_peak = peaks["bf16_tflops_sustained"] if long_region else peaks["bf16_tflops"]
-    flops_a32 = 2.0 * N_POINTS * K * DIM
+    fp8_peak = 2.0 * bf16_peak  # nominal dense e4m3 : bf16 ratio (4.5 : 2.25 PFLOP/s)
+    flops = 2.0 * N_POINTS * K * DIM
     W = (DIM + 31) // 32
     popc_aR = float(N_POINTS) * K * 4 * W
     popc_peak = SM_COUNT * POPC_PER_CLK_SM * peaks["sm_max_mhz"] * 1e6  # per second
     kernels = {
-        "assign_f32": {"ms": t_a32, "bound": "tensor", "achieved": flops_a32 / (t_a32 / 1e3) / 1e12,
+        "assign_f32": {"ms": t_a32, "bound": "tensor", "achieved": flops / (t_a32 / 1e3) / 1e12,
                        "peak": bf16_peak, "unit": "TFLOP/s",
-                       "algorithmic": f"2*N*k*d = {flops_a32:.3e} flop per launch"},
-        "assign_rbq1": {"ms": t_aR, "bound": "alu", "achieved": popc_aR / (t_aR / 1e3) / 1e12, "peak":
-                        popc_peak / 1e12, "unit": "Tpopc/s",
-                        "algorithmic": f"N*k*4*ceil(d/32) = {popc_aR:.3e} POPC per launch"},
+                       "algorithmic": f"2*N*k*d = {flops:.3e} bf16 flop per launch (screen GEMM)"},
+        "assign_rbq1": {"ms": t_aR, "bound": "tensor", "achieved": flops / (t_aR / 1e3) / 1e12,
+                        "peak": fp8_peak, "unit": "TFLOP/s",
+                        "algorithmic": f"2*N*k*d = {flops:.3e} e4m3 flop per launch (exact integer P)"},
     }
+    if t_pop is not None:
+        kernels["assign_rbq1_popcount"] = {
+            "ms": t_pop, "bound": "alu", "achieved": popc_aR / (t_pop / 1e3) / 1e12,
+            "peak": popc_peak / 1e12, "unit": "Tpopc/s", "in_step": False,
+            "algorithmic": f"N*k*4*ceil(d/32) = {popc_aR:.3e} POPC per launch"}
     for kd in kernels.values():
         kd["frac"] = kd["achieved"] / kd["peak"]
-    dom = max(kernels, key=lambda n: kernels[n]["ms"])
+    dom = max((n for n in kernels if kernels[n].get("in_step", True)), key=lambda n: kernels[n]["ms"])
     kd = kernels[dom]
     roofline = {"bound": kd["bound"], "achieved": round(kd["achieved"], 4), "peak": round(kd["peak"], 4),
                 "unit": kd["unit"], "frac": round(kd["frac"], 5), "traffic": None, "kernel": dom,
-                "peak_source": f"{peaks['source']} ({'sustained' if long_region else 'burst'} bf16)"
-                if kd["bound"] == "tensor" else f"{SM_COUNT} SMs x {POPC_PER_CLK_SM} POPC/clk x "
-                                                f"{peaks['sm_max_mhz']:.0f} MHz"}
+                "peak_source": f"{peaks['source']} ({'sustained' if long_region else 'burst'} bf16"
+                               f"{', x2 for e4m3' if dom == 'assign_rbq1' else ''})"}
 
     # ---- end to end through the C ABI with host buffers ----------------------
     e2e = None
@@ -275,8 +293,9 @@ def run_ours(args):
         Xd2 = torch.empty_like(X)
         Cd32 = torch.empty_like(C32)
         CdR = torch.empty_like(Cr)
-        pts2 = skm.Points(skm.REPR_F32, Xd2, DIM)  # screening copy rebuilt inside every call
+        pts2 = skm.Points(skm.REPR_F32, Xd2, DIM)  # screening copies rebuilt inside every call
         wsA2 = skm.workspace(skm.OP_ASSIGN, pts2, K)
+        wsAR2 = skm.workspace(skm.OP_ASSIGN, skm.rbq1_points(q, DIM, e), K)
         h2d = X_host.numel() * 4 + 2 * K * DIM * 4
         d2h = 2 * N_POINTS * 4 + 2 * K * DIM * 4
         e2e_steps = max(2, min(args.steps, 5))
@@ -293,7 +312,7 @@ def run_ours(args):
             pR2 = skm.rbq1_points(qq, DIM, e)
             skm.skm_assign(pts2, Cd32, K, want_dist=False, ws=wsA2, out=a32)
             skm.skm_update(pts2, a32, Cd32, counts=cnt32, ws=wsU32)
-            skm.skm_assign(pR2, CdR, K, want_dist=False, ws=wsAR, out=aR)
+            skm.skm_assign(pR2, CdR, K, want_dist=False, ws=wsAR2, out=aR)
             skm.skm_update(pR2, aR, CdR, counts=cntR, ws=wsUR)
             a_host[0].copy_(a32, non_blocking=True)
             a_host[1].copy_(aR, non_blocking=True)
@@ -327,7 +346,7 @@ def run_ours(args):
         line = {
             "metric": METRIC, "value": value, "unit": "distances/s", "n_gpus": world, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": ms_step, "higher_is_better": True, "scaling": "weak",
-            "vs_baseline": None, "dtype": "f32 (bf16 screen + fp32 rescore) / u32 popcount",
+            "vs_baseline": None, "dtype": "f32 (bf16 tensor screen + fp32 rescore) / 1-bit (e4m3 tensor, exact)",
             "data": "synthetic (seeded GMM embeddings, generated on the GPU)",
             "config": {"workload": WORKLOAD, "n": N_POINTS, "d": DIM, "k": K, "reprs": ["f32", "rbq1"],
                        "step": "one Lloyd iteration (assign + update) per representation",
@@ -430,8 +449,12 @@ def run_case(args):
             skm.skm_update(pts, a, C.clone(), counts=cnt, ws=wsU)
     e1.record()
     torch.cuda.synchronize()
-    print(json.dumps({"case": args.case, "n": n, "d": d, "k": k, "reps": args.reps,
-                      "ms_per_call": e0.elapsed_time(e1) / args.reps}))
+    out = {"case": args.case, "n": n, "d": d, "k": k, "reps": args.reps,
+           "ms_per_call": e0.elapsed_time(e1) / args.reps}
+    if args.case == "assign_f32":  # how often the screen alone decides a row
+        _, _, _, _, stats = skm.skm_fit(pts, k, 0, C_init=C, want_objective=False, want_dist=False)
+        out["screen_stats"] = stats
+    print(json.dumps(out))
 
 
 def main():
@@ -442,6 +465,7 @@ def main():
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-popcount", action="store_true")
     ap.add_argument("--case", default=None,
                     help="single-operation run for profiling: assign_f32|assign_rbq1|assign_sq8|update_f32|"
                          "update_rbq1|update_sq8")

@@ -6,23 +6,31 @@
 //               (bf16, 128-byte swizzle) per stage, 4-stage mbarrier ring
 //   warp 1      MMA issuer: 4 x tcgen05.mma.kind::f16 (M=128, N=256, K=16)
 //               per stage into one of two 128 x 256 fp32 TMEM accumulators
-//   warps 2-5   epilogue: tcgen05.ld of the accumulator (thread = point row),
-//               fused per-row reduction over centroids, so the N x K distance
-//               matrix never leaves the SM
+//   warps 2-9   epilogue: tcgen05.ld of the accumulator (thread = point row;
+//               two warps per TMEM lane quarter, each taking half of the 256
+//               columns), fused per-row reduction over centroids, so the
+//               N x K distance matrix never leaves the SM; the two halves of a
+//               row merge through shared memory at the end of a point tile
 // Two epilogues:
 //  SCREEN (fp32 / bf16 points): bf16 operands, so the dot product carries a
 //    rounding error.  Each pair gets a rigorous interval [L, U] for
 //    s = ||c||^2 - 2 x.c (the distance minus ||x||^2) from per-row and
-//    per-centroid bf16 residual norms.  Per row the epilogue keeps the T
-//    smallest L, the smallest U (Umin) and the smallest L it did not keep
-//    (Lev).  The nearest centroid has L <= Umin, so a row whose only such
-//    candidate is its first is decided; rows with 2..T candidates are
-//    re-scored exactly in fp32; rows with Lev <= Umin are rescanned over all
-//    k in fp32.
+//    per-centroid bf16 residual norms.  Per row the epilogue keeps the
+//    smallest U (Umin), the T smallest L among pairs with L <= Umin at the
+//    time they are seen (a pair above the running Umin can never be the
+//    nearest), and the smallest such L it could not keep (Lev).  The nearest
+//    centroid has L <= Umin, so a row whose only such candidate is its first
+//    is decided; rows with 2..T candidates are re-scored exactly in fp32;
+//    rows with Lev <= Umin are rescanned over all k in fp32.
 //  SQ8: centred codes (code - 128) are exact in bf16 and every partial sum is
 //    an integer below 2^24 for d <= 1024, so the fp32 accumulator holds the
 //    exact integer dot product; the epilogue forms the integer distance and
 //    keeps the argmin (ties to the lowest index).
+//  RBQ1: point bits as e4m3 {0, 1} and centroid SQ4 codes as e4m3 {0..15}
+//    (kind::f8f6f4, K = 32 per instruction); the accumulator holds the exact
+//    integer P = sum_i xbar_i ybar_i of Eq. final:rabitq, and the epilogue
+//    evaluates the estimator in fp32 in the library's fixed order, so the
+//    result equals the AND+popcount kernel's bit for bit.
 #include <cuda.h>
 #include <cudaTypedefs.h>
 
@@ -39,13 +47,15 @@ constexpr int BK = 64;   // bf16 elements per 128-byte swizzle row
 constexpr int STAGES = 4;
 constexpr int A_STAGE = BM * BK * 2;  // 16 KiB
 constexpr int B_STAGE = BN * BK * 2;  // 32 KiB
-constexpr int EPI_WARPS = 4;
+constexpr int EPI_WARPS = 8;  // two per TMEM lane quarter
 constexpr int THREADS = 64 + 32 * EPI_WARPS;
 constexpr int TCAND = 4;
 constexpr unsigned long long WAIT_LIMIT_NS = 2000000000ull;  // 2 s per barrier wait
-constexpr size_t SMEM_BYTES = 1024 + (size_t)STAGES * (A_STAGE + B_STAGE) + 256;
+constexpr int MERGE_WORDS = 2 * TCAND + 2;                    // one row's screen state
+constexpr int MERGE_BYTES = 2 * BM * MERGE_WORDS * 4;         // double-buffered by point tile
+constexpr size_t SMEM_BYTES = 1024 + (size_t)STAGES * (A_STAGE + B_STAGE) + 256 + MERGE_BYTES;
 
-enum { MODE_SCREEN = 0, MODE_SQ8 = 1 };
+enum { MODE_SCREEN = 0, MODE_SQ8 = 1, MODE_RBQ1 = 2 };
 
 struct TcParams {
     int64_t n;
@@ -53,7 +63,7 @@ struct TcParams {
     int k;
     int nct;  // centroid tiles
     int nkc;  // 64-wide k-slices
-    const float4 *cinfo;  // SCREEN: per centroid (||c||^2, h, ||c||, z)
+    const float4 *cinfo;  // SCREEN: per centroid (||c||^2, h', z, -), padded to 256
     const float2 *xinfo;  // SCREEN: per point (||x~||, ||x~ - x||)
     int32_t *cand;        // SCREEN: [n][TCAND + 1]
     int32_t *resc_rows;
@@ -61,8 +71,14 @@ struct TcParams {
     int32_t *counters;  // [0] rescore rows, [1] fallback rows, [2] abort flag
     int32_t *assign;
     const int32_t *nx;  // SQ8: centred ||x||^2
-    const int32_t *nc;  // SQ8: centred ||c||^2
-    float *dist;        // SQ8 (may be null)
+    const int32_t *nc;  // SQ8: centred ||c||^2, padded to 256 with a large value
+    float *dist;        // SQ8 / RBQ1 (may be null)
+    const Rbq1CInfo *rinfo;  // RBQ1: per centroid (b, s, sum ybar, ||c - m||^2), padded
+    const float *nx2;        // RBQ1 per point
+    const float *F;
+    const int32_t *popx;
+    int d;
+    float isd;  // fl(1 / sqrt(d))
 };
 
 // ------------------------------------------------------------- PTX helpers
@@ -139,6 +155,15 @@ __device__ __forceinline__ void tc_mma(uint32_t dtmem, uint64_t adesc, uint64_t 
         "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate)
         : "memory");
 }
+__device__ __forceinline__ void tc_mma_f8(uint32_t dtmem, uint64_t adesc, uint64_t bdesc,
+                                          uint32_t idesc, uint32_t accumulate) {
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "setp.ne.b32 p, %4, 0;\n\t"
+        "tcgen05.mma.cta_group::1.kind::f8f6f4 [%0], %1, %2, %3, p;\n\t}\n" ::"r"(dtmem),
+        "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate)
+        : "memory");
+}
 // 32 lanes x 32 consecutive 32-bit columns: thread i receives lane (base + i).
 __device__ __forceinline__ void tmem_ld32(uint32_t taddr, uint32_t (&v)[32]) {
     asm volatile(
@@ -167,66 +192,52 @@ __device__ __forceinline__ uint64_t sw128_desc(uint32_t saddr) {
     return d;
 }
 
-// Instruction descriptor, kind::f16: D fp32, A/B bf16, both K-major,
-// N = 256, M = 128.
+// Instruction descriptors: D fp32, both operands K-major, N = 256, M = 128;
+// kind::f16 with A/B bf16, kind::f8f6f4 with A/B e4m3.
 constexpr uint32_t IDESC = (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(BN >> 3) << 17) |
                            ((uint32_t)(BM >> 4) << 24);
+constexpr uint32_t IDESC_F8 = (1u << 4) | ((uint32_t)(BN >> 3) << 17) | ((uint32_t)(BM >> 4) << 24);
 
 // ------------------------------------------------------ screening row state
+// Per point row: the T smallest lower bounds L (sorted, indices J) among
+// centroids that could still be the nearest, the smallest upper bound Umin,
+// and Lev, the smallest such L that did not fit in the list.
 struct ScreenRow {
     float L[TCAND];
     int J[TCAND];
     float umin, lev;
-    float a, r;  // ||x~||, ||x~ - x||
 };
 
-__device__ __forceinline__ void screen_init(ScreenRow &s, float2 xi) {
+__device__ __forceinline__ void screen_init(ScreenRow &s) {
 #pragma unroll
     for (int t = 0; t < TCAND; ++t) {
         s.L[t] = INFINITY;
-        s.J[t] = -1;
+        s.J[t] = 0x7fffffff;
     }
     s.umin = INFINITY;
     s.lev = INFINITY;
-    s.a = xi.x;
-    s.r = xi.y;
 }
 
-__device__ __forceinline__ void screen_take(ScreenRow &s, float acc, float4 ci, int j) {
-    const float sv = fmaf(-2.0f, acc, ci.x);        // ||c||^2 - 2 x~.c~
-    float t = fmaf(s.a, ci.y, ci.w);                 // bound / 2
-    t = fmaf(s.r, ci.z, t);
-    const float L = fmaf(-2.0f, t, sv);
-    const float U = fmaf(2.0f, t, sv);
-    s.umin = fminf(s.umin, U);
-    if (L < s.L[TCAND - 1]) {
-        s.lev = fminf(s.lev, s.L[TCAND - 1]);
-        // insertion into the sorted list (strict <: earlier index first on ties)
-        if (L < s.L[2]) {
-            s.L[3] = s.L[2];
-            s.J[3] = s.J[2];
-            if (L < s.L[1]) {
-                s.L[2] = s.L[1];
-                s.J[2] = s.J[1];
-                if (L < s.L[0]) {
-                    s.L[1] = s.L[0];
-                    s.J[1] = s.J[0];
-                    s.L[0] = L;
-                    s.J[0] = j;
-                } else {
-                    s.L[1] = L;
-                    s.J[1] = j;
-                }
-            } else {
-                s.L[2] = L;
-                s.J[2] = j;
-            }
-        } else {
-            s.L[3] = L;
-            s.J[3] = j;
-        }
-    } else {
+// Insert (L, j) into the sorted list; what falls off the end is kept in lev.
+// (L, j) pairs are ordered by L, then by j.
+__device__ __forceinline__ void screen_insert(ScreenRow &s, float L, int j) {
+    const bool before3 = L < s.L[3] || (L == s.L[3] && j < s.J[3]);
+    if (!before3) {
         s.lev = fminf(s.lev, L);
+        return;
+    }
+    s.lev = fminf(s.lev, s.L[3]);
+    float cl = L;
+    int cj = j;
+#pragma unroll
+    for (int t = 0; t < TCAND; ++t) {  // bubble the new pair into place
+        const bool lt = cl < s.L[t] || (cl == s.L[t] && cj < s.J[t]);
+        const float tl = s.L[t];
+        const int tj = s.J[t];
+        s.L[t] = lt ? cl : tl;
+        s.J[t] = lt ? cj : tj;
+        cl = lt ? tl : cl;
+        cj = lt ? tj : cj;
     }
 }
 
@@ -247,9 +258,11 @@ __global__ void __launch_bounds__(THREADS, 1)
     auto tfull_bar = [&](int b) { return bar0 + 8u * (2 * STAGES + b); };
     auto tempty_bar = [&](int b) { return bar0 + 8u * (2 * STAGES + 2 + b); };
     uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(bars + 2 * STAGES + 4);
+    // the epilogue's merge buffer starts 256 bytes after tmem_slot (see SMEM_BYTES)
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     volatile int32_t *abort_flag = p.counters + 2;
+    constexpr int KC_ELEMS = (MODE == MODE_RBQ1) ? 128 : 64;  // elements per 128-byte row
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < STAGES; ++s) {
@@ -285,8 +298,8 @@ __global__ void __launch_bounds__(THREADS, 1)
                         const uint32_t s = it % STAGES, ph = (it / STAGES) & 1u;
                         if (!mbar_wait(empty_bar(s), ph ^ 1u, abort_flag)) goto producer_done;
                         mbar_expect_tx(full_bar(s), A_STAGE + B_STAGE);
-                        tma_load_2d(sA + s * A_STAGE, &tmA, kc * BK, (int)(rt * BM), full_bar(s));
-                        tma_load_2d(sB + s * B_STAGE, &tmB, kc * BK, ct * BN, full_bar(s));
+                        tma_load_2d(sA + s * A_STAGE, &tmA, kc * KC_ELEMS, (int)(rt * BM), full_bar(s));
+                        tma_load_2d(sB + s * B_STAGE, &tmB, kc * KC_ELEMS, ct * BN, full_bar(s));
                     }
         producer_done:;
         }
@@ -306,8 +319,12 @@ __global__ void __launch_bounds__(THREADS, 1)
                         const uint64_t ad = sw128_desc(sA + s * A_STAGE);
                         const uint64_t bd = sw128_desc(sB + s * B_STAGE);
 #pragma unroll
-                        for (int kk = 0; kk < BK / 16; ++kk)
-                            tc_mma(dcol, ad + 2u * kk, bd + 2u * kk, IDESC, (kc | kk) != 0);
+                        for (int kk = 0; kk < 4; ++kk) {  // 4 x 32-byte K steps per 128-byte row
+                            if (MODE == MODE_RBQ1)
+                                tc_mma_f8(dcol, ad + 2u * kk, bd + 2u * kk, IDESC_F8, (kc | kk) != 0);
+                            else
+                                tc_mma(dcol, ad + 2u * kk, bd + 2u * kk, IDESC, (kc | kk) != 0);
+                        }
                         tc_commit(empty_bar(s));
                     }
                     tc_commit(tfull_bar(b));
@@ -315,47 +332,96 @@ __global__ void __launch_bounds__(THREADS, 1)
         mma_done:;
         }
     } else {  // ------------------------------------------------------- epilogue
-        const int q = warp & 3;  // TMEM lane quarter this warp may access
-        const int rin = q * 32 + lane;
+        const int e = warp - 2;          // 0..7
+        const int q = warp & 3;          // TMEM lane quarter this warp may access
+        const int half = e >> 2;         // which 128 of the 256 columns
+        const int rin = q * 32 + lane;   // row within the point tile
+        uint32_t *merge = reinterpret_cast<uint32_t *>(tmem_slot + 64);  // [2][BM][MERGE_WORDS]
         uint32_t job = 0;
-        for (int64_t rt = blockIdx.x; rt < p.nrt; rt += gridDim.x) {
+        uint32_t tile = 0;
+        for (int64_t rt = blockIdx.x; rt < p.nrt; rt += gridDim.x, ++tile) {
             const int64_t row = rt * BM + rin;
             const bool valid = row < p.n;
             ScreenRow sr;
-            int32_t best = 0x7fffffff, besti = 0;
+            screen_init(sr);
+            int32_t best = 0x7fffffff, besti = 0x7fffffff;
+            float fbest = INFINITY;
+            float a2 = 0.0f, rnx2 = 0.0f, rF = 0.0f, rpc = 0.0f;
             int32_t nxr = 0;
-            if (MODE == MODE_SCREEN)
-                screen_init(sr, valid ? p.xinfo[row] : make_float2(0.f, 0.f));
-            else
+            if (MODE == MODE_SCREEN) {
+                a2 = valid ? 2.0f * p.xinfo[row].x : 0.0f;
+            } else if (MODE == MODE_SQ8) {
                 nxr = valid ? p.nx[row] : 0;
+            } else {
+                rnx2 = valid ? p.nx2[row] : 0.0f;
+                rF = valid ? p.F[row] : 0.0f;
+                rpc = valid ? (float)(2 * p.popx[row] - p.d) : 0.0f;
+            }
             for (int ct = 0; ct < p.nct; ++ct, ++job) {
                 const uint32_t b = job & 1u, bph = (job >> 1) & 1u;
                 const bool ok = mbar_wait(tfull_bar(b), bph, abort_flag);
                 if (!__all_sync(0xffffffffu, ok)) goto epi_done;
                 tc_fence_after();
-                const uint32_t taddr = tmem + ((uint32_t)(q * 32) << 16) + b * BN;
+                const uint32_t taddr = tmem + ((uint32_t)(q * 32) << 16) + b * BN + half * (BN / 2);
+                const int jh = ct * BN + half * (BN / 2);
 #pragma unroll 1
-                for (int c = 0; c < BN / 32; ++c) {
-                    const int j0 = ct * BN + c * 32;
+                for (int c = 0; c < BN / 64; ++c) {
+                    const int j0 = jh + c * 32;
                     if (j0 >= p.k) break;  // warp-uniform
                     uint32_t v[32];
                     tmem_ld32(taddr + c * 32, v);
                     if (MODE == MODE_SCREEN) {
+                        // pass 1: bounds for all 32 pairs (records are padded
+                        // with ||c||^2 = +inf, so L = U = +inf past k)
+                        float cu = INFINITY;
+#pragma unroll
+                        for (int g = 0; g < 4; ++g) {
+                            // groups of 8 loads: bounds register pressure
+                            asm volatile("" ::: "memory");
+#pragma unroll
+                            for (int i = 8 * g; i < 8 * g + 8; ++i) {
+                                const float4 ci = __ldg(p.cinfo + j0 + i);
+                                const float m = fmaf(-2.0f, __uint_as_float(v[i]), ci.x);
+                                const float w = fmaf(a2, ci.y, ci.z);
+                                cu = fminf(cu, m + w);
+                                v[i] = __float_as_uint(m - w);
+                            }
+                        }
+                        sr.umin = fminf(sr.umin, cu);
+                        // pass 2: only pairs that can still be the nearest
 #pragma unroll
                         for (int i = 0; i < 32; ++i) {
-                            const int j = j0 + i;
-                            if (j < p.k) screen_take(sr, __uint_as_float(v[i]), __ldg(p.cinfo + j), j);
+                            const float L = __uint_as_float(v[i]);
+                            if (L <= sr.umin) screen_insert(sr, L, j0 + i);
+                        }
+                    } else if (MODE == MODE_SQ8) {
+#pragma unroll
+                        for (int i = 0; i < 32; ++i) {
+                            const int32_t dot = __float2int_rn(__uint_as_float(v[i]));
+                            const int32_t dd = nxr + __ldg(p.nc + j0 + i) - 2 * dot;
+                            if (dd < best) {
+                                best = dd;
+                                besti = j0 + i;
+                            }
                         }
                     } else {
+                        // Eq. final:rabitq in Eq. rabitq_l2, fixed fp32 order
 #pragma unroll
-                        for (int i = 0; i < 32; ++i) {
-                            const int j = j0 + i;
-                            if (j < p.k) {
-                                const int32_t dot = __float2int_rn(__uint_as_float(v[i]));
-                                const int32_t dd = nxr + __ldg(p.nc + j) - 2 * dot;
-                                if (dd < best) {
-                                    best = dd;
-                                    besti = j;
+                        for (int g = 0; g < 4; ++g) {
+                            asm volatile("" ::: "memory");
+#pragma unroll
+                            for (int i = 8 * g; i < 8 * g + 8; ++i) {
+                                const float4 ci = __ldg(reinterpret_cast<const float4 *>(p.rinfo + j0 + i));
+                                const int P = __float2int_rn(__uint_as_float(v[i]));
+                                const float t1 = __fmul_rn(ci.y, __int2float_rn(2 * P - __float_as_int(ci.z)));
+                                const float t2 = __fmul_rn(ci.x, rpc);
+                                const float ip = __fmul_rn(__fadd_rn(t1, t2), p.isd);
+                                const float nn = __fadd_rn(rnx2, ci.w);
+                                const float fi = __fmul_rn(rF, ip);
+                                const float est = __fsub_rn(nn, __fmul_rn(2.0f, fi));
+                                if (est < fbest) {
+                                    fbest = est;
+                                    besti = j0 + i;
                                 }
                             }
                         }
@@ -364,28 +430,67 @@ __global__ void __launch_bounds__(THREADS, 1)
                 tc_fence_before();
                 mbar_arrive(tempty_bar(b));
             }
-            if (valid) {
+            // merge the two column halves of each row: half 1 publishes, half 0 finishes
+            uint32_t *slot = merge + ((tile & 1u) * BM + rin) * MERGE_WORDS;
+            if (half == 1) {
                 if (MODE == MODE_SCREEN) {
+#pragma unroll
+                    for (int t = 0; t < TCAND; ++t) {
+                        slot[t] = __float_as_uint(sr.L[t]);
+                        slot[TCAND + t] = (uint32_t)sr.J[t];
+                    }
+                    slot[2 * TCAND] = __float_as_uint(sr.umin);
+                    slot[2 * TCAND + 1] = __float_as_uint(sr.lev);
+                } else if (MODE == MODE_SQ8) {
+                    slot[0] = (uint32_t)best;
+                    slot[1] = (uint32_t)besti;
+                } else {
+                    slot[0] = __float_as_uint(fbest);
+                    slot[1] = (uint32_t)besti;
+                }
+            }
+            asm volatile("bar.sync 1, %0;" ::"n"(EPI_WARPS * 32) : "memory");
+            if (half == 0 && valid) {
+                if (MODE == MODE_SCREEN) {
+                    sr.umin = fminf(sr.umin, __uint_as_float(slot[2 * TCAND]));
+                    sr.lev = fminf(sr.lev, __uint_as_float(slot[2 * TCAND + 1]));
+#pragma unroll
+                    for (int t = 0; t < TCAND; ++t)
+                        screen_insert(sr, __uint_as_float(slot[t]), (int)slot[TCAND + t]);
                     int ncert = 0;
 #pragma unroll
                     for (int t = 0; t < TCAND; ++t) ncert += (sr.L[t] <= sr.umin) ? 1 : 0;
                     const bool overflow = !(sr.lev > sr.umin);
+                    const int first = sr.J[0] < p.k ? sr.J[0] : 0;
+                    p.assign[row] = first;
                     if (!overflow && ncert == 1) {
-                        p.assign[row] = sr.J[0];
+                        // decided by the screen
                     } else if (!overflow && ncert >= 2) {
                         int32_t *cr = p.cand + row * (TCAND + 1);
 #pragma unroll
                         for (int t = 0; t < TCAND; ++t) cr[t] = sr.J[t];
                         cr[TCAND] = ncert;
-                        p.assign[row] = sr.J[0];
                         p.resc_rows[atomicAdd(&p.counters[0], 1)] = (int32_t)row;
                     } else {
-                        p.assign[row] = sr.J[0] >= 0 ? sr.J[0] : 0;
                         p.fall_rows[atomicAdd(&p.counters[1], 1)] = (int32_t)row;
                     }
-                } else {
+                } else if (MODE == MODE_SQ8) {
+                    const int32_t ob = (int32_t)slot[0], oi = (int32_t)slot[1];
+                    if (ob < best || (ob == best && oi < besti)) {
+                        best = ob;
+                        besti = oi;
+                    }
                     p.assign[row] = besti;
                     if (p.dist) p.dist[row] = (float)best;
+                } else {
+                    const float ob = __uint_as_float(slot[0]);
+                    const int32_t oi = (int32_t)slot[1];
+                    if (ob < fbest || (ob == fbest && oi < besti)) {
+                        fbest = ob;
+                        besti = oi;
+                    }
+                    p.assign[row] = besti;
+                    if (p.dist) p.dist[row] = fbest;
                 }
             }
         }
@@ -405,7 +510,8 @@ __global__ void __launch_bounds__(THREADS, 1)
 // fp32 points -> bf16 screening copy (row stride dp) and per-row
 // (||x~||, ||x~ - x||), both rounded up.  One warp per row.
 __global__ void screen_prep_f32_kernel(const float *__restrict__ X, int64_t n, int d, int dp,
-                                       __nv_bfloat16 *__restrict__ xs, float2 *__restrict__ xinfo) {
+                                       __nv_bfloat16 *__restrict__ xs, float2 *__restrict__ xinfo,
+                                       unsigned int *__restrict__ rho_max_bits) {
     const int lane = threadIdx.x & 31;
     const int64_t warp = (blockIdx.x * (int64_t)blockDim.x + threadIdx.x) >> 5;
     const int64_t nw = ((int64_t)gridDim.x * blockDim.x) >> 5;
@@ -424,9 +530,14 @@ __global__ void screen_prep_f32_kernel(const float *__restrict__ X, int64_t n, i
             a2 += __shfl_xor_sync(0xffffffffu, a2, o);
             r2 += __shfl_xor_sync(0xffffffffu, r2, o);
         }
-        if (lane == 0)
-            xinfo[r] = make_float2(__double2float_ru(sqrt(a2) * (1.0 + 1e-6)),
-                                   __double2float_ru(sqrt(r2) * (1.0 + 1e-6)));
+        if (lane == 0) {
+            const float an = __double2float_ru(sqrt(a2) * (1.0 + 1e-6));
+            const float rn = __double2float_ru(sqrt(r2) * (1.0 + 1e-6));
+            xinfo[r] = make_float2(an, rn);
+            // ratio ||x~ - x|| / ||x~|| (rounded up); x~ = 0 only when x = 0
+            const float rho = an > 0.0f ? __fdiv_ru(rn, an) : 0.0f;
+            atomicMax(rho_max_bits, __float_as_uint(rho));  // non-negative: bits order as values
+        }
     }
 }
 
@@ -470,16 +581,23 @@ __global__ void screen_prep_sq8_kernel(const uint8_t *__restrict__ X, int64_t n,
     }
 }
 
-// Centroids (fp32) -> bf16 operand + (||c||^2, h, ||c||, z) with
-// h = e + (eps_acc + eps_s) (||c|| + e), e = ||c~ - c||, z = eps_s ||c||^2 / 2,
-// so that |s~ - s| <= 2 (||x~|| h + ||x~ - x|| ||c|| + z) (see the header).
-__global__ void cprep_f32_kernel(const float *__restrict__ C, int k, int d, int dp, float eps_acc,
-                                 float eps_s, __nv_bfloat16 *__restrict__ cs,
-                                 float4 *__restrict__ cinfo) {
+// Centroids (fp32) -> bf16 operand + (||c||^2, h', z, 0) with
+// h' = e + (eps_acc + eps_s) (||c|| + e) + rho_max ||c||, e = ||c~ - c||,
+// z = eps_s ||c||^2, where rho_max >= ||x~ - x|| / ||x~|| over all points, so
+// |s~ - s| <= 2 ||x~|| h' + z = w (the half-width of the pair's interval).
+// Records j in [k, kp) get ||c||^2 = +inf so they never matter.
+__global__ void cprep_f32_kernel(const float *__restrict__ C, int k, int kp, int d, int dp,
+                                 float eps_acc, float eps_s, const float *__restrict__ rho_max,
+                                 __nv_bfloat16 *__restrict__ cs, float4 *__restrict__ cinfo) {
     const int lane = threadIdx.x & 31;
     const int warp = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
     const int nw = (gridDim.x * blockDim.x) >> 5;
-    for (int j = warp; j < k; j += nw) {
+    const double rho = (double)*rho_max;
+    for (int j = warp; j < kp; j += nw) {
+        if (j >= k) {
+            if (lane == 0) cinfo[j] = make_float4(INFINITY, 0.0f, 0.0f, 0.0f);
+            continue;
+        }
         double c2 = 0.0, e2 = 0.0;
         for (int i = lane; i < d; i += 32) {
             const float c = C[(int64_t)j * d + i];
@@ -496,22 +614,26 @@ __global__ void cprep_f32_kernel(const float *__restrict__ C, int k, int d, int 
         }
         if (lane == 0) {
             const double up = 1.0 + 1e-6;
-            const double cn = sqrt(c2), e = sqrt(e2) * up;
+            const double cn = sqrt(c2) * up, e = sqrt(e2) * up;
             const double g = (cn + e) * up;
-            const double h = (e + ((double)eps_acc + (double)eps_s) * g) * up;
-            const double z = 0.5 * (double)eps_s * c2 * up;
-            cinfo[j] = make_float4(__double2float_rn(c2), __double2float_ru(h),
-                                   __double2float_ru(cn * up), __double2float_ru(z));
+            const double h = (e + ((double)eps_acc + (double)eps_s) * g + rho * cn) * up;
+            const double z = (double)eps_s * c2 * up;
+            cinfo[j] = make_float4(__double2float_rn(c2), __double2float_ru(h), __double2float_ru(z),
+                                   0.0f);
         }
     }
 }
 
-__global__ void cprep_sq8_kernel(const uint8_t *__restrict__ C, int k, int d, int dp,
+__global__ void cprep_sq8_kernel(const uint8_t *__restrict__ C, int k, int kp, int d, int dp,
                                  __nv_bfloat16 *__restrict__ cs, int32_t *__restrict__ nc) {
     const int lane = threadIdx.x & 31;
     const int warp = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
     const int nw = (gridDim.x * blockDim.x) >> 5;
-    for (int j = warp; j < k; j += nw) {
+    for (int j = warp; j < kp; j += nw) {
+        if (j >= k) {  // padding records: never the nearest
+            if (lane == 0) nc[j] = 0x3fffffff;
+            continue;
+        }
         int32_t s = 0;
         for (int i = lane; i < d; i += 32) {
             const int32_t v = (int32_t)C[(int64_t)j * d + i] - 128;
@@ -522,6 +644,48 @@ __global__ void cprep_sq8_kernel(const uint8_t *__restrict__ C, int k, int d, in
         for (int o = 16; o > 0; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
         if (lane == 0) nc[j] = s;
     }
+}
+
+// RBQ1 points: sign bits -> e4m3 bytes (bit 1 -> 1.0 = 0x38, bit 0 -> 0), row
+// stride dp bytes.  One thread per 32-bit code word writes 32 bytes.
+__global__ void screen_prep_rbq1_kernel(const uint32_t *__restrict__ codes, int64_t n, int d,
+                                        int dp, uint8_t *__restrict__ xs) {
+    const int W = (d + 31) >> 5;
+    const int64_t total = n * W;
+    for (int64_t t = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; t < total;
+         t += (int64_t)gridDim.x * blockDim.x) {
+        const int64_t r = t / W;
+        const int w = (int)(t - r * W);
+        const uint32_t bits = codes[t];
+        uint8_t *dst = xs + r * dp + 32 * w;
+        const int nb = min(32, d - 32 * w);
+        if (nb == 32 && (dp % 16) == 0) {
+            uint4 o[2];
+            uint32_t *ow = reinterpret_cast<uint32_t *>(o);
+#pragma unroll
+            for (int q = 0; q < 8; ++q) {
+                uint32_t v = 0;
+#pragma unroll
+                for (int u = 0; u < 4; ++u) v |= ((bits >> (4 * q + u)) & 1u) ? (0x38u << (8 * u)) : 0u;
+                ow[q] = v;
+            }
+            reinterpret_cast<uint4 *>(dst)[0] = o[0];
+            reinterpret_cast<uint4 *>(dst)[1] = o[1];
+        } else {
+            for (int u = 0; u < nb; ++u) dst[u] = ((bits >> u) & 1u) ? 0x38 : 0x00;
+        }
+    }
+}
+
+__global__ void pad_rbq1_info_kernel(Rbq1CInfo *__restrict__ info, int k, int kp) {
+    const int j = k + blockIdx.x * blockDim.x + threadIdx.x;
+    if (j >= kp) return;
+    Rbq1CInfo in;
+    in.b = 0.0f;
+    in.s = 0.0f;
+    in.sumy = 0;
+    in.ny2 = INFINITY;  // never the nearest
+    info[j] = in;
 }
 
 // ------------------------------------------------------------ fp32 rescoring
@@ -610,17 +774,20 @@ PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
     return fn;
 }
 
-// 2D bf16 map over [rows][cols] (row stride `stride_elems`), box = box_rows x 64.
+// 2D map over [rows][cols] of 2-byte (bf16) or 1-byte (e4m3, as uint8)
+// elements with row stride `stride_elems`; box = box_rows x 128 bytes.
 int make_map(CUtensorMap *m, const void *ptr, int64_t rows, int cols, int stride_elems,
-             int box_rows) {
+             int box_rows, int elem_bytes) {
     auto fn = encode_fn();
     if (!fn) return set_error(SKM_ERR_CUDA, "cuTensorMapEncodeTiled entry point not found");
     cuuint64_t gdim[2] = {(cuuint64_t)cols, (cuuint64_t)rows};
-    cuuint64_t gstride[1] = {(cuuint64_t)stride_elems * 2};
-    cuuint32_t box[2] = {(cuuint32_t)BK, (cuuint32_t)box_rows};
+    cuuint64_t gstride[1] = {(cuuint64_t)stride_elems * elem_bytes};
+    cuuint32_t box[2] = {(cuuint32_t)(128 / elem_bytes), (cuuint32_t)box_rows};
     cuuint32_t estr[2] = {1, 1};
-    CUresult r = fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void *>(ptr), gdim, gstride,
-                    box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+    const CUtensorMapDataType dt =
+        elem_bytes == 2 ? CU_TENSOR_MAP_DATA_TYPE_BFLOAT16 : CU_TENSOR_MAP_DATA_TYPE_UINT8;
+    CUresult r = fn(m, dt, 2, const_cast<void *>(ptr), gdim, gstride, box, estr,
+                    CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
                     CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
     if (r != CUDA_SUCCESS) return set_error(SKM_ERR_CUDA, "cuTensorMapEncodeTiled failed (%d)", (int)r);
     return SKM_OK;
@@ -636,8 +803,8 @@ int device_sms() {
 template <int MODE>
 int launch_tc(const void *xs, int64_t n, int dp, int d, const void *cs, int k, const TcParams &p0,
               cudaStream_t st) {
-    static std::once_flag attr_once[2];
-    static cudaError_t attr_err[2] = {cudaSuccess, cudaSuccess};
+    static std::once_flag attr_once[3];
+    static cudaError_t attr_err[3] = {cudaSuccess, cudaSuccess, cudaSuccess};
     std::call_once(attr_once[MODE], [] {
         attr_err[MODE] = cudaFuncSetAttribute(tc_assign_kernel<MODE>,
                                               cudaFuncAttributeMaxDynamicSharedMemorySize,
@@ -646,14 +813,15 @@ int launch_tc(const void *xs, int64_t n, int dp, int d, const void *cs, int k, c
     if (attr_err[MODE] != cudaSuccess)
         return set_error(SKM_ERR_CUDA, "cudaFuncSetAttribute: %s", cudaGetErrorString(attr_err[MODE]));
     CUtensorMap ma, mb;
-    SKM_TRY(make_map(&ma, xs, n, d, dp, BM));
-    SKM_TRY(make_map(&mb, cs, k, d, dp, BN));
+    const int eb = MODE == MODE_RBQ1 ? 1 : 2;
+    SKM_TRY(make_map(&ma, xs, n, d, dp, BM, eb));
+    SKM_TRY(make_map(&mb, cs, k, d, dp, BN, eb));
     TcParams p = p0;
     p.n = n;
     p.nrt = cdiv(n, BM);
     p.k = k;
     p.nct = (int)cdiv(k, BN);
-    p.nkc = (int)cdiv(d, BK);
+    p.nkc = (int)cdiv(d, 128 / eb);
     const int grid = (int)std::min<int64_t>(device_sms(), p.nrt);
     tc_assign_kernel<MODE><<<grid, THREADS, SMEM_BYTES, st>>>(ma, mb, p);
     SKM_CUDA_TRY(launched());
@@ -667,6 +835,7 @@ int grid_warps(int64_t items) {
 }
 
 inline int round8(int d) { return (d + 7) & ~7; }
+inline int round16(int d) { return (d + 15) & ~15; }
 
 }  // namespace
 
@@ -678,6 +847,7 @@ size_t tc_screen_bytes(int repr, int64_t n, int d, const void *x) {
     case SKM_REPR_F32:
         cv.take<uint16_t>((size_t)n * dp);
         cv.take<float2>(n);
+        cv.take<float>(1);
         break;
     case SKM_REPR_SQ8:
         if (d > TC_SQ8_MAX_D) return 0;
@@ -687,6 +857,10 @@ size_t tc_screen_bytes(int repr, int64_t n, int d, const void *x) {
     case SKM_REPR_BF16:
         if (d % 8 != 0 || ((uintptr_t)x & 15) != 0) cv.take<uint16_t>((size_t)n * dp);
         cv.take<float2>(n);
+        cv.take<float>(1);
+        break;
+    case SKM_REPR_RBQ1:
+        cv.take<uint8_t>((size_t)n * round16(d));
         break;
     default:
         return 0;
@@ -697,6 +871,7 @@ size_t tc_screen_bytes(int repr, int64_t n, int d, const void *x) {
 struct ScreenView {
     const void *xs = nullptr;
     const float2 *xinfo = nullptr;
+    const float *rho_max = nullptr;  // max over points of ||x~ - x|| / ||x~||
     const int32_t *nx = nullptr;
 };
 
@@ -708,6 +883,7 @@ static ScreenView screen_view(int repr, int64_t n, int d, const void *x, const v
     case SKM_REPR_F32:
         v.xs = cv.take<uint16_t>((size_t)n * dp);
         v.xinfo = cv.take<float2>(n);
+        v.rho_max = cv.take<float>(1);
         break;
     case SKM_REPR_SQ8:
         v.xs = cv.take<uint16_t>((size_t)n * dp);
@@ -719,6 +895,10 @@ static ScreenView screen_view(int repr, int64_t n, int d, const void *x, const v
         else
             v.xs = x;
         v.xinfo = cv.take<float2>(n);
+        v.rho_max = cv.take<float>(1);
+        break;
+    case SKM_REPR_RBQ1:
+        v.xs = cv.take<uint8_t>((size_t)n * round16(d));
         break;
     }
     return v;
@@ -729,10 +909,12 @@ int tc_screen_prep(const skm_data *x, void *screen, cudaStream_t st) {
     const int d = x->d, dp = round8(d);
     ScreenView v = screen_view(x->repr, n, d, x->x, screen);
     const int g = grid_warps(n);
+    if (v.rho_max) SKM_CUDA_TRY(cudaMemsetAsync((void *)v.rho_max, 0, sizeof(float), st));
     switch (x->repr) {
     case SKM_REPR_F32:
         screen_prep_f32_kernel<<<g, 256, 0, st>>>(static_cast<const float *>(x->x), n, d, dp,
-                                                  (__nv_bfloat16 *)v.xs, (float2 *)v.xinfo);
+                                                  (__nv_bfloat16 *)v.xs, (float2 *)v.xinfo,
+                                                  (unsigned int *)v.rho_max);
         break;
     case SKM_REPR_SQ8:
         screen_prep_sq8_kernel<<<g, 256, 0, st>>>(static_cast<const uint8_t *>(x->x), n, d, dp,
@@ -743,6 +925,13 @@ int tc_screen_prep(const skm_data *x, void *screen, cudaStream_t st) {
                                                    v.xs == x->x ? nullptr : (uint16_t *)v.xs,
                                                    (float2 *)v.xinfo);
         break;
+    case SKM_REPR_RBQ1: {
+        int64_t blocks = (n * words_of(d) + 255) / 256;
+        if (blocks > 152 * 8) blocks = 152 * 8;
+        screen_prep_rbq1_kernel<<<(int)blocks, 256, 0, st>>>(static_cast<const uint32_t *>(x->x), n,
+                                                             d, round16(d), (uint8_t *)v.xs);
+        break;
+    }
     default:
         return set_error(SKM_ERR_INVALID_ARG, "no screening copy for repr %d", x->repr);
     }
@@ -755,18 +944,24 @@ void tc_plan(int repr, int64_t n, int d, int k, const void *x, const void *scree
     b.stats = cv.take<int64_t>(4);
     b.counters = cv.take<int32_t>(4);
     const int dp = round8(d);
-    const bool dense = repr == SKM_REPR_F32 || repr == SKM_REPR_BF16 ||
+    const bool dense = repr == SKM_REPR_F32 || repr == SKM_REPR_BF16 || repr == SKM_REPR_RBQ1 ||
                        (repr == SKM_REPR_SQ8 && d <= TC_SQ8_MAX_D);
     if (!dense) return;
     if (!screen) {
         const size_t sb = tc_screen_bytes(repr, n, d, x);
         b.screen = cv.take<uint8_t>(sb);
     }
+    const size_t kp = (size_t)cdiv(k, BN) * BN;  // per-centroid records padded to whole tiles
+    if (repr == SKM_REPR_RBQ1) {
+        b.cs = reinterpret_cast<uint16_t *>(cv.take<uint8_t>((size_t)k * round16(d)));
+        b.rinfo = cv.take<Rbq1CInfo>(kp);
+        return;
+    }
     b.cs = cv.take<uint16_t>((size_t)k * dp);
     if (repr == SKM_REPR_SQ8) {
-        b.nc = cv.take<int32_t>(k);
+        b.nc = cv.take<int32_t>(kp);
     } else {
-        b.cinfo = cv.take<float4>(k);
+        b.cinfo = cv.take<float4>(kp);
         b.cand = cv.take<int32_t>((size_t)n * (TCAND + 1));
         b.resc_rows = cv.take<int32_t>(n);
         b.fall_rows = cv.take<int32_t>(n);
@@ -793,8 +988,9 @@ int tc_assign_float(const skm_data *x, const float *C, int k, int32_t *assign, f
     const int nkc = (int)cdiv(d, BK);
     const float eps_acc = (float)((nkc * (BK / 16) + 4) * 0x1p-18);
     const float eps_s = 0x1p-21f;
-    cprep_f32_kernel<<<grid_warps(k), 256, 0, st>>>(C, k, d, dp, eps_acc, eps_s,
-                                                    (__nv_bfloat16 *)b.cs, b.cinfo);
+    const int kp = (int)(cdiv(k, BN) * BN);
+    cprep_f32_kernel<<<grid_warps(kp), 256, 0, st>>>(C, k, kp, d, dp, eps_acc, eps_s, v.rho_max,
+                                                     (__nv_bfloat16 *)b.cs, b.cinfo);
     SKM_CUDA_TRY(launched());
     SKM_CUDA_TRY(cudaMemsetAsync(b.counters, 0, sizeof(int32_t) * 4, st));
     TcParams p{};
@@ -852,7 +1048,8 @@ int tc_assign_sq8(const skm_data *x, const uint8_t *C, int k, int32_t *nx_plain,
         screen = b.screen;
     }
     ScreenView v = screen_view(x->repr, n, d, x->x, screen);
-    cprep_sq8_kernel<<<grid_warps(k), 256, 0, st>>>(C, k, d, dp, (__nv_bfloat16 *)b.cs, b.nc);
+    const int kp = (int)(cdiv(k, BN) * BN);
+    cprep_sq8_kernel<<<grid_warps(kp), 256, 0, st>>>(C, k, kp, d, dp, (__nv_bfloat16 *)b.cs, b.nc);
     SKM_CUDA_TRY(launched());
     SKM_CUDA_TRY(cudaMemsetAsync(b.counters, 0, sizeof(int32_t) * 4, st));
     TcParams p{};
@@ -862,6 +1059,41 @@ int tc_assign_sq8(const skm_data *x, const uint8_t *C, int k, int32_t *nx_plain,
     p.nc = b.nc;
     p.dist = dist;
     SKM_TRY(launch_tc<MODE_SQ8>(v.xs, n, dp, d, b.cs, k, p, st));
+    add_stats_kernel<<<1, 1, 0, st>>>(b.counters, b.stats);
+    SKM_CUDA_TRY(launched());
+    return SKM_OK;
+}
+
+int tc_assign_rbq1(const skm_data *x, const float *C, int k, int32_t *assign, float *dist,
+                   TcAssignBufs &b, cudaStream_t st) {
+    const int64_t n = x->n;
+    const int d = x->d, dp = round16(d);
+    const void *screen = x->screen;
+    if (!screen) {
+        skm_data tmp = *x;
+        SKM_TRY(tc_screen_prep(&tmp, b.screen, st));
+        screen = b.screen;
+    }
+    ScreenView v = screen_view(x->repr, n, d, x->x, screen);
+    const int kp = (int)(cdiv(k, BN) * BN);
+    SKM_CUDA_TRY(launch_rbq1_cprep_tc(C, k, d, x->m, reinterpret_cast<uint8_t *>(b.cs), dp, b.rinfo,
+                                      st));
+    if (kp > k) {
+        pad_rbq1_info_kernel<<<(kp - k + 255) / 256, 256, 0, st>>>(b.rinfo, k, kp);
+        SKM_CUDA_TRY(launched());
+    }
+    SKM_CUDA_TRY(cudaMemsetAsync(b.counters, 0, sizeof(int32_t) * 4, st));
+    TcParams p{};
+    p.counters = b.counters;
+    p.assign = assign;
+    p.dist = dist;
+    p.rinfo = b.rinfo;
+    p.nx2 = x->nx2;
+    p.F = x->F;
+    p.popx = x->popx;
+    p.d = d;
+    p.isd = (float)(1.0 / sqrt((double)d));
+    SKM_TRY(launch_tc<MODE_RBQ1>(v.xs, n, dp, d, b.cs, k, p, st));
     add_stats_kernel<<<1, 1, 0, st>>>(b.counters, b.stats);
     SKM_CUDA_TRY(launched());
     return SKM_OK;

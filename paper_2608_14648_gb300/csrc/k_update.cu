@@ -114,48 +114,97 @@ cudaError_t launch_scatter(const int32_t *assign, int64_t n, int k, const int64_
 }
 
 // ------------------------------------------------------ segmented sums: float
-// One CTA per cluster; thread t owns dimensions t, t + 256, ... (up to 16).
-// Members are read four at a time for memory-level parallelism.
-constexpr int SEG_THREADS = 256;
-constexpr int SEG_MAXV = 16;  // d <= 4096
+// One CTA per cluster, 8 warps; warp w takes members w, w + 8, ... (two rows
+// in flight), lane l accumulates 16-byte column groups l, l + 32, ... of a
+// 1024-element column chunk.  Warp partials meet in shared memory and are
+// summed in warp order.
+constexpr int SEG_WARPS = 8;
+constexpr int SEG_THREADS = SEG_WARPS * 32;
+constexpr int SEG_CHUNK = 1024;  // columns per pass (float: 8 float4 per lane)
+
+template <bool BF16>
+__device__ __forceinline__ void seg_load8(const void *X, int64_t p, int d, int c0, int lane,
+                                          float (&v)[SEG_CHUNK / 32]) {
+    // columns c0 + 4*(lane + 32*g) .. +3 for g = 0..7 (zero past d)
+#pragma unroll
+    for (int g = 0; g < SEG_CHUNK / 128; ++g) {
+        const int c = c0 + 4 * (lane + 32 * g);
+        float4 f = make_float4(0.f, 0.f, 0.f, 0.f);
+        if (BF16) {
+            const uint16_t *x = reinterpret_cast<const uint16_t *>(X) + p * d;
+            if (c + 3 < d && (d % 4) == 0) {
+                const uint2 w = __ldg(reinterpret_cast<const uint2 *>(x + c));
+                f = make_float4(__uint_as_float(w.x << 16), __uint_as_float(w.x & 0xffff0000u),
+                                __uint_as_float(w.y << 16), __uint_as_float(w.y & 0xffff0000u));
+            } else {
+                float t[4];
+#pragma unroll
+                for (int u = 0; u < 4; ++u)
+                    t[u] = (c + u < d) ? __uint_as_float(((uint32_t)__ldg(x + c + u)) << 16) : 0.f;
+                f = make_float4(t[0], t[1], t[2], t[3]);
+            }
+        } else {
+            const float *x = reinterpret_cast<const float *>(X) + p * d;
+            if (c + 3 < d && (d % 4) == 0) {
+                f = __ldg(reinterpret_cast<const float4 *>(x + c));
+            } else {
+                float t[4];
+#pragma unroll
+                for (int u = 0; u < 4; ++u) t[u] = (c + u < d) ? __ldg(x + c + u) : 0.f;
+                f = make_float4(t[0], t[1], t[2], t[3]);
+            }
+        }
+        v[4 * g] = f.x;
+        v[4 * g + 1] = f.y;
+        v[4 * g + 2] = f.z;
+        v[4 * g + 3] = f.w;
+    }
+}
 
 template <bool BF16>
 __global__ void __launch_bounds__(SEG_THREADS) segsum_float_kernel(
     const void *__restrict__ Xv, int d, const int32_t *__restrict__ perm,
     const int64_t *__restrict__ offsets, float *__restrict__ C, double *__restrict__ partial) {
+    __shared__ float red[SEG_WARPS][SEG_CHUNK];
     const int j = blockIdx.x;
     const int64_t lo = offsets[j], hi = offsets[j + 1];
     const int64_t cnt = hi - lo;
     if (cnt == 0) return;  // empty cluster keeps its centroid / adds nothing
-    float acc[SEG_MAXV];
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    for (int c0 = 0; c0 < d; c0 += SEG_CHUNK) {
+        float acc[SEG_CHUNK / 32];
 #pragma unroll
-    for (int v = 0; v < SEG_MAXV; ++v) acc[v] = 0.0f;
-    for (int64_t q = lo; q < hi; ++q) {
-        const int64_t p = perm[q];
-        if (BF16) {
-            const uint16_t *x = reinterpret_cast<const uint16_t *>(Xv) + p * d;
+        for (int t = 0; t < SEG_CHUNK / 32; ++t) acc[t] = 0.0f;
+        int64_t q = lo + warp;
+        for (; q + SEG_WARPS < hi; q += 2 * SEG_WARPS) {
+            float v0[SEG_CHUNK / 32], v1[SEG_CHUNK / 32];
+            seg_load8<BF16>(Xv, perm[q], d, c0, lane, v0);
+            seg_load8<BF16>(Xv, perm[q + SEG_WARPS], d, c0, lane, v1);
 #pragma unroll
-            for (int v = 0; v < SEG_MAXV; ++v) {
-                const int i = threadIdx.x + v * SEG_THREADS;
-                if (i < d) acc[v] += __uint_as_float(((uint32_t)__ldg(x + i)) << 16);
-            }
-        } else {
-            const float *x = reinterpret_cast<const float *>(Xv) + p * d;
-#pragma unroll
-            for (int v = 0; v < SEG_MAXV; ++v) {
-                const int i = threadIdx.x + v * SEG_THREADS;
-                if (i < d) acc[v] += __ldg(x + i);
-            }
+            for (int t = 0; t < SEG_CHUNK / 32; ++t) acc[t] += v0[t] + v1[t];
         }
-    }
+        if (q < hi) {
+            float v0[SEG_CHUNK / 32];
+            seg_load8<BF16>(Xv, perm[q], d, c0, lane, v0);
 #pragma unroll
-    for (int v = 0; v < SEG_MAXV; ++v) {
-        const int i = threadIdx.x + v * SEG_THREADS;
-        if (i < d) {
+            for (int t = 0; t < SEG_CHUNK / 32; ++t) acc[t] += v0[t];
+        }
+        __syncthreads();
+#pragma unroll
+        for (int g = 0; g < SEG_CHUNK / 128; ++g)
+#pragma unroll
+            for (int u = 0; u < 4; ++u) red[warp][4 * (lane + 32 * g) + u] = acc[4 * g + u];
+        __syncthreads();
+        for (int t = threadIdx.x; t < SEG_CHUNK; t += SEG_THREADS) {
+            const int i = c0 + t;
+            if (i >= d) break;
+            float s = 0.0f;
+#pragma unroll
+            for (int w = 0; w < SEG_WARPS; ++w) s += red[w][t];
             if (partial)
-                partial[(int64_t)j * d + i] += (double)acc[v];
+                partial[(int64_t)j * d + i] += (double)s;
             else
-                C[(int64_t)j * d + i] = __fdiv_rn(acc[v], (float)cnt);
+                C[(int64_t)j * d + i] = __fdiv_rn(s, (float)cnt);
         }
     }
 }
@@ -179,33 +228,60 @@ __device__ __forceinline__ uint8_t round_half_even_div(int64_t S, int64_t m) {
     return (uint8_t)q;
 }
 
+// Warp w takes members w, w + 8, ...; lane l sums bytes 4l..4l+3 of each
+// 128-byte column group; exact integer partials are combined with shared
+// memory atomics (order-independent).
 __global__ void __launch_bounds__(SEG_THREADS) segsum_sq8_kernel(
     const uint8_t *__restrict__ X, int d, const int32_t *__restrict__ perm,
     const int64_t *__restrict__ offsets, uint8_t *__restrict__ C, int64_t *__restrict__ partial) {
+    __shared__ unsigned long long tot[SEG_CHUNK];
     const int j = blockIdx.x;
     const int64_t lo = offsets[j], hi = offsets[j + 1];
     const int64_t cnt = hi - lo;
     if (cnt == 0) return;
-    int64_t acc[SEG_MAXV];
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const bool vec = (d % 4) == 0;
+    for (int c0 = 0; c0 < d; c0 += SEG_CHUNK) {
+        for (int t = threadIdx.x; t < SEG_CHUNK; t += SEG_THREADS) tot[t] = 0ull;
+        __syncthreads();
+        uint32_t acc[SEG_CHUNK / 32];  // columns c0 + 4*(lane + 32 g) + u
 #pragma unroll
-    for (int v = 0; v < SEG_MAXV; ++v) acc[v] = 0;
-    for (int64_t q = lo; q < hi; ++q) {
-        const uint8_t *x = X + (int64_t)perm[q] * d;
+        for (int t = 0; t < SEG_CHUNK / 32; ++t) acc[t] = 0u;
+        for (int64_t q = lo + warp; q < hi; q += SEG_WARPS) {
+            const uint8_t *x = X + (int64_t)perm[q] * d;
 #pragma unroll
-        for (int v = 0; v < SEG_MAXV; ++v) {
-            const int i = threadIdx.x + v * SEG_THREADS;
-            if (i < d) acc[v] += __ldg(x + i);
+            for (int g = 0; g < SEG_CHUNK / 128; ++g) {
+                const int c = c0 + 4 * (lane + 32 * g);
+                uint32_t w = 0;
+                if (vec && c + 3 < d) {
+                    w = __ldg(reinterpret_cast<const uint32_t *>(x + c));
+                } else {
+#pragma unroll
+                    for (int u = 0; u < 4; ++u)
+                        if (c + u < d) w |= ((uint32_t)__ldg(x + c + u)) << (8 * u);
+                }
+#pragma unroll
+                for (int u = 0; u < 4; ++u) acc[4 * g + u] += (w >> (8 * u)) & 0xffu;
+            }
         }
-    }
 #pragma unroll
-    for (int v = 0; v < SEG_MAXV; ++v) {
-        const int i = threadIdx.x + v * SEG_THREADS;
-        if (i < d) {
+        for (int g = 0; g < SEG_CHUNK / 128; ++g)
+#pragma unroll
+            for (int u = 0; u < 4; ++u) {
+                const int t = 4 * (lane + 32 * g) + u;
+                if (c0 + t < d && acc[4 * g + u]) atomicAdd(&tot[t], (unsigned long long)acc[4 * g + u]);
+            }
+        __syncthreads();
+        for (int t = threadIdx.x; t < SEG_CHUNK; t += SEG_THREADS) {
+            const int i = c0 + t;
+            if (i >= d) break;
+            const int64_t S = (int64_t)tot[t];
             if (partial)
-                partial[(int64_t)j * d + i] += acc[v];
+                partial[(int64_t)j * d + i] += S;
             else
-                C[(int64_t)j * d + i] = round_half_even_div(acc[v], cnt);
+                C[(int64_t)j * d + i] = round_half_even_div(S, cnt);
         }
+        __syncthreads();
     }
 }
 
@@ -229,47 +305,64 @@ __device__ __forceinline__ float rbq1_finish(int64_t T, int64_t U, int64_t cnt, 
     return __double2float_rn(__dadd_rn((double)m, v));
 }
 
+// Warp w takes members w, w + 8, ...; word t of a member is loaded by lane t
+// and broadcast; lane l owns dimension 32 t + l of every word t.  Per-warp
+// int64 partials are combined with shared-memory atomics (exact).
+constexpr int RB_WORDS = 32;  // words per pass (1024 dimensions)
+
 __global__ void __launch_bounds__(SEG_THREADS) segsum_rbq1_kernel(
     const uint32_t *__restrict__ codes, const float *__restrict__ F, int d,
     const float *__restrict__ m, int e, const int32_t *__restrict__ perm,
     const int64_t *__restrict__ offsets, float *__restrict__ C, int64_t *__restrict__ partial) {
+    __shared__ unsigned long long tot[RB_WORDS * 32];
+    __shared__ unsigned long long utot;
     const int j = blockIdx.x;
     const int64_t lo = offsets[j], hi = offsets[j + 1];
     const int64_t cnt = hi - lo;
     if (cnt == 0) return;
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int W = (d + 31) >> 5;
     const double pow2 = ldexp(1.0, e);
-    int64_t acc[SEG_MAXV];
-#pragma unroll
-    for (int v = 0; v < SEG_MAXV; ++v) acc[v] = 0;
-    int64_t U = 0;
-    for (int64_t q = lo; q < hi; ++q) {
-        const int64_t p = perm[q];
-        const int64_t fq = __double2ll_rn(__dmul_rn((double)__ldg(F + p), pow2));
-        U += fq;
-        const uint32_t *cw = codes + p * W;
-#pragma unroll
-        for (int v = 0; v < SEG_MAXV; ++v) {
-            const int i = threadIdx.x + v * SEG_THREADS;
-            if (i < d) {
-                const uint32_t word = __ldg(cw + (i >> 5));
-                if ((word >> (i & 31)) & 1u) acc[v] += fq;
-            }
-        }
-    }
     const double pow2m = ldexp(1.0, -e);
     const double isd = __ddiv_rn(1.0, __dsqrt_rn((double)d));
+    for (int w0 = 0; w0 < W; w0 += RB_WORDS) {
+        const int nw = min(RB_WORDS, W - w0);
+        for (int t = threadIdx.x; t < RB_WORDS * 32; t += SEG_THREADS) tot[t] = 0ull;
+        if (threadIdx.x == 0 && w0 == 0) utot = 0ull;  // U is summed in the first pass only
+        __syncthreads();
+        int64_t acc[RB_WORDS];
 #pragma unroll
-    for (int v = 0; v < SEG_MAXV; ++v) {
-        const int i = threadIdx.x + v * SEG_THREADS;
-        if (i < d) {
-            if (partial)
-                partial[(int64_t)j * (d + 1) + i] += acc[v];
-            else
-                C[(int64_t)j * d + i] = rbq1_finish(acc[v], U, cnt, m[i], pow2m, isd);
+        for (int t = 0; t < RB_WORDS; ++t) acc[t] = 0;
+        int64_t usum = 0;
+        for (int64_t q = lo + warp; q < hi; q += SEG_WARPS) {
+            const int64_t p = perm[q];
+            const int64_t fq = __double2ll_rn(__dmul_rn((double)__ldg(F + p), pow2));
+            usum += fq;
+            const uint32_t mine = (lane < nw) ? __ldg(codes + p * W + w0 + lane) : 0u;
+#pragma unroll
+            for (int t = 0; t < RB_WORDS; ++t) {
+                const uint32_t word = __shfl_sync(0xffffffffu, mine, t);
+                if ((word >> lane) & 1u) acc[t] += fq;
+            }
         }
+#pragma unroll
+        for (int t = 0; t < RB_WORDS; ++t)
+            if (t < nw && acc[t]) atomicAdd(&tot[32 * t + lane], (unsigned long long)acc[t]);
+        if (lane == 0 && w0 == 0) atomicAdd(&utot, (unsigned long long)usum);
+        __syncthreads();
+        const int64_t U = (int64_t)utot;
+        for (int t = threadIdx.x; t < nw * 32; t += SEG_THREADS) {
+            const int i = 32 * w0 + t;
+            if (i >= d) continue;
+            const int64_t T = (int64_t)tot[t];
+            if (partial)
+                partial[(int64_t)j * (d + 1) + i] += T;
+            else
+                C[(int64_t)j * d + i] = rbq1_finish(T, U, cnt, m[i], pow2m, isd);
+        }
+        if (partial && w0 == 0 && threadIdx.x == 0) partial[(int64_t)j * (d + 1) + d] += U;
+        __syncthreads();
     }
-    if (partial && threadIdx.x == 0) partial[(int64_t)j * (d + 1) + d] += U;
 }
 
 cudaError_t launch_segsum_rbq1(const uint32_t *codes, const float *F, int d, const float *m,

@@ -84,6 +84,8 @@ cudaError_t launch_rbq1_exponent(const float *F, int64_t n, unsigned int *maxbit
 // centroid preparation
 cudaError_t launch_rbq1_cprep(const float *C, int k, int d, const float *m, uint4 *planes,
                               Rbq1CInfo *info, cudaStream_t st);
+cudaError_t launch_rbq1_cprep_tc(const float *C, int k, int d, const float *m, uint8_t *yq, int dq,
+                                 Rbq1CInfo *info, cudaStream_t st);
 cudaError_t launch_row_sqnorm_u8(const uint8_t *codes, int64_t n, int d, int32_t *out,
                                  cudaStream_t st);
 // assignment

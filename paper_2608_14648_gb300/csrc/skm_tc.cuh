@@ -16,6 +16,7 @@ struct TcAssignBufs {
     uint16_t *cs = nullptr;       // centroid operand, bf16 [k][round8(d)]
     float4 *cinfo = nullptr;      // F32/BF16: per-centroid bound terms
     int32_t *nc = nullptr;        // SQ8: centred ||c||^2
+    Rbq1CInfo *rinfo = nullptr;   // RBQ1: per-centroid estimator terms (padded)
     int32_t *cand = nullptr;      // F32/BF16: [n][5] screen candidates + count
     int32_t *resc_rows = nullptr;
     int32_t *fall_rows = nullptr;
@@ -32,6 +33,10 @@ int tc_assign_float(const skm_data *x, const float *C, int k, int32_t *assign, f
 int tc_assign_sq8(const skm_data *x, const uint8_t *C, int k, int32_t *nx_plain,
                   int32_t *nc_plain, int32_t *assign, float *dist, TcAssignBufs &b,
                   cudaStream_t st);
+// RBQ1 on tensor cores (e4m3 operands, exact integer P, same fp32 epilogue
+// as the AND+popcount kernel).
+int tc_assign_rbq1(const skm_data *x, const float *C, int k, int32_t *assign, float *dist,
+                   TcAssignBufs &b, cudaStream_t st);
 // Copies the cumulative statistics; returns SKM_ERR_TIMEOUT if a pipeline
 // wait gave up.  Synchronises the stream.
 int tc_read_stats(const TcAssignBufs &b, skm_stats *st_host, cudaStream_t st);
