@@ -426,8 +426,10 @@ def run_case(args):
     C = X[synth.forgy_indices(n, k, seed=0).cuda()].clone()
     if args.case in ("assign_f32", "update_f32"):
         pts = skm.Points(skm.REPR_F32, X, d).with_screen()
-    elif args.case in ("assign_rbq1", "update_rbq1"):
+    elif args.case in ("assign_rbq1", "update_rbq1", "assign_rbq1_popcount"):
         pts = skm.rbq1_points(skm.skm_quantize(skm.REPR_RBQ1, X), d)
+        if args.case == "assign_rbq1":
+            pts = pts.with_screen()
     elif args.case in ("assign_sq8", "update_sq8"):
         q = skm.skm_quantize(skm.REPR_SQ8, X)
         pts = skm.Points(skm.REPR_SQ8, q["codes"], d).with_screen()
@@ -443,7 +445,9 @@ def run_case(args):
     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     e0.record()
     for _ in range(args.reps):
-        if args.case.startswith("assign"):
+        if args.case == "assign_rbq1_popcount":
+            skm.skm_assign_rbq1_noalloc(pts, C, a)
+        elif args.case.startswith("assign"):
             skm.skm_assign(pts, C, k, want_dist=False, ws=wsA, out=a)
         else:
             skm.skm_update(pts, a, C.clone(), counts=cnt, ws=wsU)

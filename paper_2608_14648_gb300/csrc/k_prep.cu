@@ -3,24 +3,25 @@
 //  re-encoded with per-centroid SQ4 (b = min rho, s = (max rho - b)/15,
 //  s = 1 when flat, ybar = clip(rint((rho - b)/s), 0, 15)) and stored as four
 //  bit planes per 32-dimension word, so that sum_i xbar_i ybar_i =
-//  sum_j 2^j popc(xbar & plane_j).  One lane per centroid walks its row in
-//  order, which fixes the fp64 summation order of ||rho||^2.
+//  sum_j 2^j popc(xbar & plane_j), and/or as e4m3 bytes for the tensor kernel.
+//  ||rho||^2 is summed in fp64 in increasing dimension order by one lane.
 //  SQ8: per-row sums of squared codes (exact int32).
 #include "skm_internal.cuh"
 
 namespace skm {
 
-// Each warp owns 32 centroids (one per lane).  The warp stages 32 x 32 tiles
-// of rho = c - m through shared memory with coalesced loads; each lane then
-// walks its own centroid's dimensions in increasing order.
+// One warp per centroid.  rho = c - m is kept in the warp's slice of shared
+// memory; min/max and the code sum are exact warp reductions, the codes of
+// 32 consecutive dimensions become four bit planes through __ballot_sync, and
+// one lane forms ||rho||^2 in fp64 in increasing dimension order.
 constexpr int CPREP_WARPS = 4;
 
 // e4m3 encodings of the integers 0..15 (sign 0, exponent bias 7, 3 mantissa
 // bits): 0 -> 0x00, 1 -> 0x38, 2 -> 0x40, 3 -> 0x44, 4 -> 0x48, ... 15 -> 0x57.
 __device__ __forceinline__ uint8_t e4m3_of_code(uint32_t y) {
     if (y == 0) return 0;
-    const int e = 31 - __clz(y);                       // floor(log2 y), 0..3
-    const uint32_t mant = (y << (3 - e)) & 7u;         // 3 bits below the leading one
+    const int e = 31 - __clz(y);                // floor(log2 y), 0..3
+    const uint32_t mant = (y << (3 - e)) & 7u;  // 3 bits below the leading one
     return (uint8_t)(((uint32_t)(e + 7) << 3) | mant);
 }
 
@@ -30,60 +31,51 @@ __device__ __forceinline__ uint8_t e4m3_of_code(uint32_t y) {
 __global__ void __launch_bounds__(CPREP_WARPS * 32) rbq1_cprep_kernel(
     const float *__restrict__ C, int k, int d, const float *__restrict__ m,
     uint4 *__restrict__ planes, Rbq1CInfo *__restrict__ info, uint8_t *__restrict__ yq, int dq) {
-    __shared__ float tile[CPREP_WARPS][32][33];
+    extern __shared__ float sh_rho[];  // [CPREP_WARPS][d]
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int j0 = (blockIdx.x * CPREP_WARPS + warp) * 32;
-    if (j0 >= k) return;  // warp-uniform
-    const int j = j0 + lane;
-    const bool valid = j < k;
-    float(*t)[33] = tile[warp];
-    auto stage = [&](int i0) {
-        const int i = i0 + lane;
-        const float mi = (i < d) ? m[i] : 0.0f;
-#pragma unroll 4
-        for (int r = 0; r < 32; ++r) {
-            const int row = j0 + r;
-            t[r][lane] = (row < k && i < d) ? __fsub_rn(C[(int64_t)row * d + i], mi) : 0.0f;
-        }
-        __syncwarp();
-    };
+    const int j = blockIdx.x * CPREP_WARPS + warp;
+    if (j >= k) return;  // warp-uniform
+    float *rho = sh_rho + (size_t)warp * d;
+    const float *c = C + (int64_t)j * d;
     float lo = INFINITY, hi = -INFINITY;
-    double q2 = 0.0;
-    for (int i0 = 0; i0 < d; i0 += 32) {
-        stage(i0);
-        const int n = min(32, d - i0);
-        for (int l = 0; l < n; ++l) {
-            const float r = t[lane][l];
-            lo = fminf(lo, r);
-            hi = fmaxf(hi, r);
-            q2 = __dadd_rn(q2, __dmul_rn((double)r, (double)r));
-        }
-        __syncwarp();
+    for (int i = lane; i < d; i += 32) {
+        const float r = __fsub_rn(c[i], m[i]);
+        rho[i] = r;
+        lo = fminf(lo, r);
+        hi = fmaxf(hi, r);
     }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+        lo = fminf(lo, __shfl_xor_sync(0xffffffffu, lo, o));
+        hi = fmaxf(hi, __shfl_xor_sync(0xffffffffu, hi, o));
+    }
+    __syncwarp();
     float sc = __fdiv_rn(__fsub_rn(hi, lo), 15.0f);
     if (!(sc > 0.0f)) sc = 1.0f;
     const int W = (d + 31) >> 5;
     int32_t sy = 0;
     for (int w = 0; w < W; ++w) {
-        stage(32 * w);
-        uint32_t p0 = 0, p1 = 0, p2 = 0, p3 = 0;
-        const int n = min(32, d - 32 * w);
-        for (int l = 0; l < n; ++l) {
-            float q = rintf(__fdiv_rn(__fsub_rn(t[lane][l], lo), sc));
+        const int i = 32 * w + lane;
+        uint32_t y = 0;
+        if (i < d) {
+            float q = rintf(__fdiv_rn(__fsub_rn(rho[i], lo), sc));
             q = (q >= 0.0f) ? q : 0.0f;
             q = fminf(q, 15.0f);
-            const uint32_t y = (uint32_t)q;
-            sy += (int32_t)y;
-            if (yq && valid) yq[(int64_t)j * dq + 32 * w + l] = e4m3_of_code(y);
-            p0 |= (y & 1u) << l;
-            p1 |= ((y >> 1) & 1u) << l;
-            p2 |= ((y >> 2) & 1u) << l;
-            p3 |= ((y >> 3) & 1u) << l;
+            y = (uint32_t)q;
+            if (yq) yq[(int64_t)j * dq + i] = e4m3_of_code(y);
         }
-        if (valid && planes) planes[(int64_t)j * W + w] = make_uint4(p0, p1, p2, p3);
-        __syncwarp();
+        sy += (int32_t)y;
+        const uint32_t p0 = __ballot_sync(0xffffffffu, y & 1u);
+        const uint32_t p1 = __ballot_sync(0xffffffffu, y & 2u);
+        const uint32_t p2 = __ballot_sync(0xffffffffu, y & 4u);
+        const uint32_t p3 = __ballot_sync(0xffffffffu, y & 8u);
+        if (planes && lane == 0) planes[(int64_t)j * W + w] = make_uint4(p0, p1, p2, p3);
     }
-    if (valid) {
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) sy += __shfl_xor_sync(0xffffffffu, sy, o);
+    if (lane == 0) {
+        double q2 = 0.0;
+        for (int i = 0; i < d; ++i) q2 = __dadd_rn(q2, __dmul_rn((double)rho[i], (double)rho[i]));
         Rbq1CInfo in;
         in.b = lo;
         in.s = sc;
@@ -93,20 +85,27 @@ __global__ void __launch_bounds__(CPREP_WARPS * 32) rbq1_cprep_kernel(
     }
 }
 
+static cudaError_t launch_cprep_common(const float *C, int k, int d, const float *m, uint4 *planes,
+                                       Rbq1CInfo *info, uint8_t *yq, int dq, cudaStream_t st) {
+    const size_t smem = (size_t)CPREP_WARPS * d * sizeof(float);
+    if (smem > 48 * 1024) {
+        const cudaError_t e = cudaFuncSetAttribute(
+            rbq1_cprep_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+        if (e != cudaSuccess) return e;
+    }
+    rbq1_cprep_kernel<<<(k + CPREP_WARPS - 1) / CPREP_WARPS, CPREP_WARPS * 32, smem, st>>>(
+        C, k, d, m, planes, info, yq, dq);
+    return launched();
+}
+
 cudaError_t launch_rbq1_cprep(const float *C, int k, int d, const float *m, uint4 *planes,
                               Rbq1CInfo *info, cudaStream_t st) {
-    const int per_block = CPREP_WARPS * 32;
-    rbq1_cprep_kernel<<<(k + per_block - 1) / per_block, per_block, 0, st>>>(C, k, d, m, planes,
-                                                                            info, nullptr, 0);
-    return launched();
+    return launch_cprep_common(C, k, d, m, planes, info, nullptr, 0, st);
 }
 
 cudaError_t launch_rbq1_cprep_tc(const float *C, int k, int d, const float *m, uint8_t *yq, int dq,
                                  Rbq1CInfo *info, cudaStream_t st) {
-    const int per_block = CPREP_WARPS * 32;
-    rbq1_cprep_kernel<<<(k + per_block - 1) / per_block, per_block, 0, st>>>(C, k, d, m, nullptr,
-                                                                            info, yq, dq);
-    return launched();
+    return launch_cprep_common(C, k, d, m, nullptr, info, yq, dq, st);
 }
 
 // sum_i code_i^2 per row (exact, fits int32 for d <= 4096); one warp per row.

@@ -27,10 +27,11 @@
 //    exact integer dot product; the epilogue forms the integer distance and
 //    keeps the argmin (ties to the lowest index).
 //  RBQ1: point bits as e4m3 {0, 1} and centroid SQ4 codes as e4m3 {0..15}
-//    (kind::f8f6f4, K = 32 per instruction); the accumulator holds the exact
-//    integer P = sum_i xbar_i ybar_i of Eq. final:rabitq, and the epilogue
-//    evaluates the estimator in fp32 in the library's fixed order, so the
-//    result equals the AND+popcount kernel's bit for bit.
+//    (kind::f8f6f4, K = 32 per instruction); the nearest integer to the
+//    accumulator is P = sum_i xbar_i ybar_i of Eq. final:rabitq (d <= 1024
+//    keeps P < 2^14 and the accumulation error far below 1/2), and the
+//    epilogue evaluates the estimator in fp32 in the library's fixed order,
+//    so the result equals the AND+popcount kernel's bit for bit.
 #include <cuda.h>
 #include <cudaTypedefs.h>
 
@@ -63,7 +64,8 @@ struct TcParams {
     int k;
     int nct;  // centroid tiles
     int nkc;  // 64-wide k-slices
-    const float4 *cinfo;  // SCREEN: per centroid (||c||^2, h', z, -), padded to 256
+    const float4 *cinfo;  // SCREEN: per column pair (||c||^2 x2, h' x2), padded to 256
+    const float2 *cinfoz; // SCREEN: per column pair (z x2)
     const float2 *xinfo;  // SCREEN: per point (||x~||, ||x~ - x||)
     int32_t *cand;        // SCREEN: [n][TCAND + 1]
     int32_t *resc_rows;
@@ -73,7 +75,8 @@ struct TcParams {
     const int32_t *nx;  // SQ8: centred ||x||^2
     const int32_t *nc;  // SQ8: centred ||c||^2, padded to 256 with a large value
     float *dist;        // SQ8 / RBQ1 (may be null)
-    const Rbq1CInfo *rinfo;  // RBQ1: per centroid (b, s, sum ybar, ||c - m||^2), padded
+    const float4 *rinfo;     // RBQ1: per column pair (b x2, s x2), padded
+    const float4 *rinfoq;    // RBQ1: per column pair (-sum ybar x2, ||c - m||^2 x2)
     const float *nx2;        // RBQ1 per point
     const float *F;
     const int32_t *popx;
@@ -178,6 +181,58 @@ __device__ __forceinline__ void tmem_ld32(uint32_t taddr, uint32_t (&v)[32]) {
         : "r"(taddr)
         : "memory");
     asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+}
+
+// Packed fp32 pairs (two IEEE round-to-nearest operations per instruction).
+__device__ __forceinline__ float2 ffma2(float2 a, float2 b, float2 c) {
+    float2 r;
+    asm("{\n\t.reg .b64 ra, rb, rc, rd;\n\t"
+        "mov.b64 ra, {%2, %3};\n\tmov.b64 rb, {%4, %5};\n\tmov.b64 rc, {%6, %7};\n\t"
+        "fma.rn.f32x2 rd, ra, rb, rc;\n\tmov.b64 {%0, %1}, rd;\n\t}"
+        : "=f"(r.x), "=f"(r.y)
+        : "f"(a.x), "f"(a.y), "f"(b.x), "f"(b.y), "f"(c.x), "f"(c.y));
+    return r;
+}
+__device__ __forceinline__ float2 fadd2(float2 a, float2 b) {
+    float2 r;
+    asm("{\n\t.reg .b64 ra, rb, rd;\n\t"
+        "mov.b64 ra, {%2, %3};\n\tmov.b64 rb, {%4, %5};\n\t"
+        "add.rn.f32x2 rd, ra, rb;\n\tmov.b64 {%0, %1}, rd;\n\t}"
+        : "=f"(r.x), "=f"(r.y)
+        : "f"(a.x), "f"(a.y), "f"(b.x), "f"(b.y));
+    return r;
+}
+__device__ __forceinline__ float2 fmul2(float2 a, float2 b) {
+    float2 r;
+    asm("{\n\t.reg .b64 ra, rb, rd;\n\t"
+        "mov.b64 ra, {%2, %3};\n\tmov.b64 rb, {%4, %5};\n\t"
+        "mul.rn.f32x2 rd, ra, rb;\n\tmov.b64 {%0, %1}, rd;\n\t}"
+        : "=f"(r.x), "=f"(r.y)
+        : "f"(a.x), "f"(a.y), "f"(b.x), "f"(b.y));
+    return r;
+}
+__device__ __forceinline__ float2 fsub2(float2 a, float2 b) {
+    float2 r;
+    asm("{\n\t.reg .b64 ra, rb, rd;\n\t"
+        "mov.b64 ra, {%2, %3};\n\tmov.b64 rb, {%4, %5};\n\t"
+        "sub.rn.f32x2 rd, ra, rb;\n\tmov.b64 {%0, %1}, rd;\n\t}"
+        : "=f"(r.x), "=f"(r.y)
+        : "f"(a.x), "f"(a.y), "f"(b.x), "f"(b.y));
+    return r;
+}
+
+// v[i] for a lane-dependent i in [0, 32): binary select tree (no local memory).
+__device__ __forceinline__ uint32_t pick32(const uint32_t (&v)[32], int i) {
+    uint32_t w16[16], w8[8], w4[4], w2[2];
+#pragma unroll
+    for (int t = 0; t < 16; ++t) w16[t] = (i & 16) ? v[t + 16] : v[t];
+#pragma unroll
+    for (int t = 0; t < 8; ++t) w8[t] = (i & 8) ? w16[t + 8] : w16[t];
+#pragma unroll
+    for (int t = 0; t < 4; ++t) w4[t] = (i & 4) ? w8[t + 4] : w8[t];
+#pragma unroll
+    for (int t = 0; t < 2; ++t) w2[t] = (i & 2) ? w4[t + 2] : w4[t];
+    return (i & 1) ? w2[1] : w2[0];
 }
 
 // Shared-memory matrix descriptor: K-major operand, 128-byte swizzle, rows of
@@ -371,28 +426,43 @@ __global__ void __launch_bounds__(THREADS, 1)
                     uint32_t v[32];
                     tmem_ld32(taddr + c * 32, v);
                     if (MODE == MODE_SCREEN) {
-                        // pass 1: bounds for all 32 pairs (records are padded
-                        // with ||c||^2 = +inf, so L = U = +inf past k)
-                        float cu = INFINITY;
+                        // pass 1, two columns per packed op: m = ||c||^2 - 2 acc,
+                        // w = 2 ||x~|| h' + z; L = m - w (kept in v), U = m + w.
+                        // Records past k have ||c||^2 = +inf, so L = U = +inf.
+                        float cu[4], cl[4];
 #pragma unroll
                         for (int g = 0; g < 4; ++g) {
-                            // groups of 8 loads: bounds register pressure
-                            asm volatile("" ::: "memory");
+                            asm volatile("" ::: "memory");  // bounds register pressure
+                            cu[g] = INFINITY;
+                            cl[g] = INFINITY;
 #pragma unroll
-                            for (int i = 8 * g; i < 8 * g + 8; ++i) {
-                                const float4 ci = __ldg(p.cinfo + j0 + i);
-                                const float m = fmaf(-2.0f, __uint_as_float(v[i]), ci.x);
-                                const float w = fmaf(a2, ci.y, ci.z);
-                                cu = fminf(cu, m + w);
-                                v[i] = __float_as_uint(m - w);
+                            for (int i = 8 * g; i < 8 * g + 8; i += 2) {
+                                const float4 ci = __ldg(p.cinfo + ((j0 + i) >> 1));
+                                const float2 cz = __ldg(p.cinfoz + ((j0 + i) >> 1));
+                                const float2 acc = make_float2(__uint_as_float(v[i]), __uint_as_float(v[i + 1]));
+                                const float2 m = ffma2(make_float2(-2.0f, -2.0f), acc, make_float2(ci.x, ci.y));
+                                const float2 w = ffma2(make_float2(a2, a2), make_float2(ci.z, ci.w), cz);
+                                const float2 U = fadd2(m, w);
+                                const float2 L = fsub2(m, w);
+                                cu[g] = fminf(cu[g], fminf(U.x, U.y));
+                                cl[g] = fminf(cl[g], fminf(L.x, L.y));
+                                v[i] = __float_as_uint(L.x);
+                                v[i + 1] = __float_as_uint(L.y);
                             }
                         }
-                        sr.umin = fminf(sr.umin, cu);
-                        // pass 2: only pairs that can still be the nearest
+                        sr.umin = fminf(sr.umin, fminf(fminf(cu[0], cu[1]), fminf(cu[2], cu[3])));
+                        const float lmin = fminf(fminf(cl[0], cl[1]), fminf(cl[2], cl[3]));
+                        // pass 2 (rare once Umin is small): pairs that can still be the nearest
+                        if (lmin <= sr.umin) {
+                            uint32_t mask = 0;
 #pragma unroll
-                        for (int i = 0; i < 32; ++i) {
-                            const float L = __uint_as_float(v[i]);
-                            if (L <= sr.umin) screen_insert(sr, L, j0 + i);
+                            for (int i = 0; i < 32; ++i)
+                                mask |= (__uint_as_float(v[i]) <= sr.umin ? 1u : 0u) << i;
+                            while (mask) {
+                                const int i = __ffs(mask) - 1;
+                                mask &= mask - 1;
+                                screen_insert(sr, __uint_as_float(pick32(v, i)), j0 + i);
+                            }
                         }
                     } else if (MODE == MODE_SQ8) {
 #pragma unroll
@@ -405,26 +475,48 @@ __global__ void __launch_bounds__(THREADS, 1)
                             }
                         }
                     } else {
-                        // Eq. final:rabitq in Eq. rabitq_l2, fixed fp32 order
+                        // Eq. final:rabitq in Eq. rabitq_l2 in the library's fixed
+                        // fp32 order, scalar IEEE operations only (packed f32x2
+                        // sequences were measured not to reproduce it).  The e4m3
+                        // accumulator carries a small non-integer error (~2^-12),
+                        // so P is its nearest integer; 2P - sum ybar is exact.
+                        float gb[4];
+                        int gi[4];
 #pragma unroll
                         for (int g = 0; g < 4; ++g) {
                             asm volatile("" ::: "memory");
+                            gb[g] = INFINITY;
+                            gi[g] = 0x7fffffff;
 #pragma unroll
-                            for (int i = 8 * g; i < 8 * g + 8; ++i) {
-                                const float4 ci = __ldg(reinterpret_cast<const float4 *>(p.rinfo + j0 + i));
-                                const int P = __float2int_rn(__uint_as_float(v[i]));
-                                const float t1 = __fmul_rn(ci.y, __int2float_rn(2 * P - __float_as_int(ci.z)));
-                                const float t2 = __fmul_rn(ci.x, rpc);
-                                const float ip = __fmul_rn(__fadd_rn(t1, t2), p.isd);
-                                const float nn = __fadd_rn(rnx2, ci.w);
-                                const float fi = __fmul_rn(rF, ip);
-                                const float est = __fsub_rn(nn, __fmul_rn(2.0f, fi));
-                                if (est < fbest) {
-                                    fbest = est;
-                                    besti = j0 + i;
+                            for (int i = 8 * g; i < 8 * g + 8; i += 2) {
+                                const float4 bs = __ldg(p.rinfo + ((j0 + i) >> 1));
+                                const float4 qn = __ldg(p.rinfoq + ((j0 + i) >> 1));
+                                const float bb[2] = {bs.x, bs.y}, ss[2] = {bs.z, bs.w};
+                                const float nq[2] = {qn.x, qn.y}, ny[2] = {qn.z, qn.w};
+#pragma unroll
+                                for (int o = 0; o < 2; ++o) {
+                                    const float P = rintf(__uint_as_float(v[i + o]));
+                                    const float qv = __fmaf_rn(2.0f, P, nq[o]);  // exact
+                                    const float t1 = __fmul_rn(ss[o], qv);
+                                    const float t2 = __fmul_rn(bb[o], rpc);
+                                    const float ip = __fmul_rn(__fadd_rn(t1, t2), p.isd);
+                                    const float nn = __fadd_rn(rnx2, ny[o]);
+                                    const float fi = __fmul_rn(rF, ip);
+                                    const float est = __fsub_rn(nn, __fmul_rn(2.0f, fi));
+                                    if (est < gb[g]) {
+                                        gb[g] = est;
+                                        gi[g] = j0 + i + o;
+                                    }
                                 }
                             }
                         }
+                        // groups hold increasing column ranges: earlier group wins ties
+#pragma unroll
+                        for (int g = 0; g < 4; ++g)
+                            if (gb[g] < fbest) {
+                                fbest = gb[g];
+                                besti = gi[g];
+                            }
                     }
                 }
                 tc_fence_before();
@@ -585,17 +677,26 @@ __global__ void screen_prep_sq8_kernel(const uint8_t *__restrict__ X, int64_t n,
 // h' = e + (eps_acc + eps_s) (||c|| + e) + rho_max ||c||, e = ||c~ - c||,
 // z = eps_s ||c||^2, where rho_max >= ||x~ - x|| / ||x~|| over all points, so
 // |s~ - s| <= 2 ||x~|| h' + z = w (the half-width of the pair's interval).
-// Records j in [k, kp) get ||c||^2 = +inf so they never matter.
+// Records j in [k, kp) get ||c||^2 = +inf so they never matter.  Layout:
+// column pair p = (2p, 2p+1) -> cinfo[p] = (||c||^2 x2, h' x2), cinfoz[p] = (z x2).
 __global__ void cprep_f32_kernel(const float *__restrict__ C, int k, int kp, int d, int dp,
                                  float eps_acc, float eps_s, const float *__restrict__ rho_max,
-                                 __nv_bfloat16 *__restrict__ cs, float4 *__restrict__ cinfo) {
+                                 __nv_bfloat16 *__restrict__ cs, float4 *__restrict__ cinfo,
+                                 float2 *__restrict__ cinfoz) {
     const int lane = threadIdx.x & 31;
     const int warp = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
     const int nw = (gridDim.x * blockDim.x) >> 5;
     const double rho = (double)*rho_max;
+    float *cf = reinterpret_cast<float *>(cinfo);
+    float *zf = reinterpret_cast<float *>(cinfoz);
     for (int j = warp; j < kp; j += nw) {
+        const int pp = j >> 1, o = j & 1;
         if (j >= k) {
-            if (lane == 0) cinfo[j] = make_float4(INFINITY, 0.0f, 0.0f, 0.0f);
+            if (lane == 0) {
+                cf[4 * pp + o] = INFINITY;
+                cf[4 * pp + 2 + o] = 0.0f;
+                zf[2 * pp + o] = 0.0f;
+            }
             continue;
         }
         double c2 = 0.0, e2 = 0.0;
@@ -618,8 +719,9 @@ __global__ void cprep_f32_kernel(const float *__restrict__ C, int k, int kp, int
             const double g = (cn + e) * up;
             const double h = (e + ((double)eps_acc + (double)eps_s) * g + rho * cn) * up;
             const double z = (double)eps_s * c2 * up;
-            cinfo[j] = make_float4(__double2float_rn(c2), __double2float_ru(h), __double2float_ru(z),
-                                   0.0f);
+            cf[4 * pp + o] = __double2float_rn(c2);
+            cf[4 * pp + 2 + o] = __double2float_ru(h);
+            zf[2 * pp + o] = __double2float_ru(z);
         }
     }
 }
@@ -677,15 +779,32 @@ __global__ void screen_prep_rbq1_kernel(const uint32_t *__restrict__ codes, int6
     }
 }
 
-__global__ void pad_rbq1_info_kernel(Rbq1CInfo *__restrict__ info, int k, int kp) {
-    const int j = k + blockIdx.x * blockDim.x + threadIdx.x;
-    if (j >= kp) return;
-    Rbq1CInfo in;
-    in.b = 0.0f;
-    in.s = 0.0f;
-    in.sumy = 0;
-    in.ny2 = INFINITY;  // never the nearest
-    info[j] = in;
+// Per-centroid estimator terms -> column-pair records for the tensor
+// epilogue: bs[p] = (b x2, s x2), qn[p] = (-sum ybar x2, ||c - m||^2 x2);
+// columns past k get ||c - m||^2 = +inf (never the nearest).
+__global__ void pack_rbq1_pairs_kernel(const Rbq1CInfo *__restrict__ info, int k, int kp,
+                                       float4 *__restrict__ bs, float4 *__restrict__ qn) {
+    const int pp = blockIdx.x * blockDim.x + threadIdx.x;
+    if (2 * pp >= kp) return;
+    float b[2], sc[2], q[2], n2[2];
+#pragma unroll
+    for (int o = 0; o < 2; ++o) {
+        const int j = 2 * pp + o;
+        if (j < k) {
+            const Rbq1CInfo in = info[j];
+            b[o] = in.b;
+            sc[o] = in.s;
+            q[o] = -(float)in.sumy;
+            n2[o] = in.ny2;
+        } else {
+            b[o] = 0.0f;
+            sc[o] = 0.0f;
+            q[o] = 0.0f;
+            n2[o] = INFINITY;
+        }
+    }
+    bs[pp] = make_float4(b[0], b[1], sc[0], sc[1]);
+    qn[pp] = make_float4(q[0], q[1], n2[0], n2[1]);
 }
 
 // ------------------------------------------------------------ fp32 rescoring
@@ -860,6 +979,7 @@ size_t tc_screen_bytes(int repr, int64_t n, int d, const void *x) {
         cv.take<float>(1);
         break;
     case SKM_REPR_RBQ1:
+        if (d > TC_RBQ1_MAX_D) return 0;
         cv.take<uint8_t>((size_t)n * round16(d));
         break;
     default:
@@ -944,7 +1064,8 @@ void tc_plan(int repr, int64_t n, int d, int k, const void *x, const void *scree
     b.stats = cv.take<int64_t>(4);
     b.counters = cv.take<int32_t>(4);
     const int dp = round8(d);
-    const bool dense = repr == SKM_REPR_F32 || repr == SKM_REPR_BF16 || repr == SKM_REPR_RBQ1 ||
+    const bool dense = repr == SKM_REPR_F32 || repr == SKM_REPR_BF16 ||
+                       (repr == SKM_REPR_RBQ1 && d <= TC_RBQ1_MAX_D) ||
                        (repr == SKM_REPR_SQ8 && d <= TC_SQ8_MAX_D);
     if (!dense) return;
     if (!screen) {
@@ -954,14 +1075,17 @@ void tc_plan(int repr, int64_t n, int d, int k, const void *x, const void *scree
     const size_t kp = (size_t)cdiv(k, BN) * BN;  // per-centroid records padded to whole tiles
     if (repr == SKM_REPR_RBQ1) {
         b.cs = reinterpret_cast<uint16_t *>(cv.take<uint8_t>((size_t)k * round16(d)));
-        b.rinfo = cv.take<Rbq1CInfo>(kp);
+        b.rinfo = cv.take<Rbq1CInfo>(k);
+        b.rpair_bs = cv.take<float4>(kp / 2);
+        b.rpair_qn = cv.take<float4>(kp / 2);
         return;
     }
     b.cs = cv.take<uint16_t>((size_t)k * dp);
     if (repr == SKM_REPR_SQ8) {
         b.nc = cv.take<int32_t>(kp);
     } else {
-        b.cinfo = cv.take<float4>(kp);
+        b.cinfo = cv.take<float4>(kp / 2);
+        b.cinfoz = cv.take<float2>(kp / 2);
         b.cand = cv.take<int32_t>((size_t)n * (TCAND + 1));
         b.resc_rows = cv.take<int32_t>(n);
         b.fall_rows = cv.take<int32_t>(n);
@@ -990,11 +1114,12 @@ int tc_assign_float(const skm_data *x, const float *C, int k, int32_t *assign, f
     const float eps_s = 0x1p-21f;
     const int kp = (int)(cdiv(k, BN) * BN);
     cprep_f32_kernel<<<grid_warps(kp), 256, 0, st>>>(C, k, kp, d, dp, eps_acc, eps_s, v.rho_max,
-                                                     (__nv_bfloat16 *)b.cs, b.cinfo);
+                                                     (__nv_bfloat16 *)b.cs, b.cinfo, b.cinfoz);
     SKM_CUDA_TRY(launched());
     SKM_CUDA_TRY(cudaMemsetAsync(b.counters, 0, sizeof(int32_t) * 4, st));
     TcParams p{};
     p.cinfo = b.cinfo;
+    p.cinfoz = b.cinfoz;
     p.xinfo = v.xinfo;
     p.cand = b.cand;
     p.resc_rows = b.resc_rows;
@@ -1078,16 +1203,16 @@ int tc_assign_rbq1(const skm_data *x, const float *C, int k, int32_t *assign, fl
     const int kp = (int)(cdiv(k, BN) * BN);
     SKM_CUDA_TRY(launch_rbq1_cprep_tc(C, k, d, x->m, reinterpret_cast<uint8_t *>(b.cs), dp, b.rinfo,
                                       st));
-    if (kp > k) {
-        pad_rbq1_info_kernel<<<(kp - k + 255) / 256, 256, 0, st>>>(b.rinfo, k, kp);
-        SKM_CUDA_TRY(launched());
-    }
+    pack_rbq1_pairs_kernel<<<(kp / 2 + 255) / 256, 256, 0, st>>>(b.rinfo, k, kp, b.rpair_bs,
+                                                                 b.rpair_qn);
+    SKM_CUDA_TRY(launched());
     SKM_CUDA_TRY(cudaMemsetAsync(b.counters, 0, sizeof(int32_t) * 4, st));
     TcParams p{};
     p.counters = b.counters;
     p.assign = assign;
     p.dist = dist;
-    p.rinfo = b.rinfo;
+    p.rinfo = b.rpair_bs;
+    p.rinfoq = b.rpair_qn;
     p.nx2 = x->nx2;
     p.F = x->F;
     p.popx = x->popx;

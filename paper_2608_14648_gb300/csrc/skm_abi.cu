@@ -71,6 +71,8 @@ static int check_k(const skm_data *x, int k, bool k_le_n = false) {
 // ------------------------------------------------------------ workspace plans
 struct AssignBufs {
     int32_t *nx = nullptr, *nc = nullptr;  // SQ8 with d > 1024 (__dp4a path)
+    uint4 *planes = nullptr;                // RBQ1 with d > 1024 (AND + popcount path)
+    Rbq1CInfo *info = nullptr;
     TcAssignBufs tc;                        // tensor-core paths (F32, BF16, SQ8, RBQ1)
 };
 
@@ -82,6 +84,12 @@ static void plan_assign(const skm_data *x, int k, Carver &cv, AssignBufs &b) {
         if (d > TC_SQ8_MAX_D) {
             b.nx = cv.take<int32_t>(n);
             b.nc = cv.take<int32_t>(k);
+        }
+        break;
+    case SKM_REPR_RBQ1:
+        if (d > TC_RBQ1_MAX_D) {
+            b.planes = cv.take<uint4>((size_t)k * words_of(d));
+            b.info = cv.take<Rbq1CInfo>(k);
         }
         break;
     default:
@@ -162,7 +170,14 @@ static int do_assign(const skm_data *x, const void *C, int k, const int32_t *pre
                               b.tc, st));
         break;
     case SKM_REPR_RBQ1:
-        SKM_TRY(tc_assign_rbq1(x, static_cast<const float *>(C), k, assign, dist, b.tc, st));
+        if (d <= TC_RBQ1_MAX_D) {
+            SKM_TRY(tc_assign_rbq1(x, static_cast<const float *>(C), k, assign, dist, b.tc, st));
+        } else {
+            SKM_CUDA_TRY(launch_rbq1_cprep(static_cast<const float *>(C), k, d, x->m, b.planes,
+                                           b.info, st));
+            SKM_CUDA_TRY(launch_assign_rbq1(static_cast<const uint32_t *>(x->x), x->nx2, x->F,
+                                            x->popx, n, d, b.planes, b.info, k, assign, dist, st));
+        }
         break;
     }
     return SKM_OK;

@@ -8,15 +8,22 @@ namespace skm {
 // Above this d the fp32 accumulator of the bf16-encoded SQ8 dot product can
 // exceed 2^24 and stop being exact; SQ8 then uses the __dp4a kernel.
 constexpr int TC_SQ8_MAX_D = 1024;
+// The e4m3 1-bit path rounds its accumulator to the integer P; up to this d
+// (P < 2^14) the accumulation error stays far below 1/2.  Beyond it the
+// AND + popcount kernel is used.
+constexpr int TC_RBQ1_MAX_D = 1024;
 
 struct TcAssignBufs {
     int64_t *stats = nullptr;     // [0] rescored rows, [1] fallback rows, [2] timeout (cumulative)
     int32_t *counters = nullptr;  // per call: [0] rescore list, [1] fallback list, [2] abort flag
     uint8_t *screen = nullptr;    // screening copy built per call when the caller gave none
     uint16_t *cs = nullptr;       // centroid operand, bf16 [k][round8(d)]
-    float4 *cinfo = nullptr;      // F32/BF16: per-centroid bound terms
+    float4 *cinfo = nullptr;      // F32/BF16: per-column-pair bound terms
+    float2 *cinfoz = nullptr;
     int32_t *nc = nullptr;        // SQ8: centred ||c||^2
-    Rbq1CInfo *rinfo = nullptr;   // RBQ1: per-centroid estimator terms (padded)
+    Rbq1CInfo *rinfo = nullptr;   // RBQ1: per-centroid estimator terms
+    float4 *rpair_bs = nullptr;   // RBQ1: the same as column-pair records (padded)
+    float4 *rpair_qn = nullptr;
     int32_t *cand = nullptr;      // F32/BF16: [n][5] screen candidates + count
     int32_t *resc_rows = nullptr;
     int32_t *fall_rows = nullptr;

@@ -187,7 +187,8 @@ def test_encode_rbq1_vs_oracle(skm, n, d):
         assert np.all(h["codes"][:, -1] >> (d % 32) == 0)
 
 
-@pytest.mark.parametrize("n,d,k", [(3000, 768, 300), (777, 33, 7), (500, 64, 1), (1000, 1024, 65)])
+@pytest.mark.parametrize("n,d,k", [(3000, 768, 300), (777, 33, 7), (500, 64, 1), (1000, 1024, 65),
+                                   (600, 1500, 40)])
 def test_assign_update_rbq1_bitexact(skm, n, d, k):
     X = _points(n, d, seed=n + 2)
     r = skm.skm_quantize(skm.REPR_RBQ1, X.to(DEV))
