@@ -59,6 +59,16 @@ typedef enum skm_repr {
 
 typedef enum skm_dtype { SKM_DTYPE_F32 = 0, SKM_DTYPE_BF16 = 1 } skm_dtype;
 
+/* skm_data.flags */
+enum {
+    /* F32 / BF16, d <= 1024: assign by exact dimension pruning on CUDA cores
+     * (Section 3.1 "SuperKMeans": partial distances over 32-dimension prefix
+     * blocks, a centroid is dropped as soon as its partial distance exceeds
+     * the row's current best) instead of the tensor-core screen.  Same
+     * result (the fp32 nearest centroid). */
+    SKM_FLAG_PRUNE = 1
+};
+
 /* Points being clustered.  Which fields are read depends on repr. */
 typedef struct skm_data {
     int32_t repr;       /* skm_repr                                          */
@@ -72,7 +82,7 @@ typedef struct skm_data {
     const float *m;     /* centring mean m               [d]                 */
     int32_t rbq1_exp;   /* fixed-point exponent e of the decode-average
                            (skm_rbq1_exponent); fit() computes it itself     */
-    int32_t reserved0;
+    int32_t flags;      /* SKM_FLAG_* (0 = defaults)                          */
     /* Optional screening copy for F32 / BF16 / SQ8 assignment, built once by
      * skm_screen_prep (the points never change across Lloyd iterations).
      * NULL: skm_assign builds it in its workspace on every call.            */
@@ -85,7 +95,10 @@ typedef struct skm_stats {
     int64_t rescored_rows;    /* F32/BF16: rows whose screen was not decisive */
     int64_t fallback_rows;    /* F32/BF16: rows rescanned over all k in fp32  */
     int64_t empty_clusters;   /* after the last update                         */
-    int64_t reserved[5];
+    int64_t prune_first_block;/* SKM_FLAG_PRUNE: (row, centroid) pairs alive
+                                 after the first 32-dimension block             */
+    int64_t prune_complete;   /* ... alive after the last block                 */
+    int64_t reserved[3];
 } skm_stats;
 
 const char *skm_last_error(void);
@@ -184,9 +197,10 @@ int skm_screen_prep(const skm_data *x, void *screen, size_t screen_bytes, void *
  *        rescoring (direct differences) of every centroid the bound cannot
  *        rule out, and an fp32 scan over all k for rows the screen could not
  *        narrow down.  dist = fp32 sum of squared differences.
- *   BF16 float [k][d] centroids against bf16 points; exact dimension
- *        pruning over 32-dimension prefix blocks (a centroid is dropped as
- *        soon as its partial distance exceeds the row's current best).
+ *   BF16 float [k][d] centroids against bf16 points (the projected points
+ *        stored in bf16): the tensor-core screen as for F32 (the bf16
+ *        points are the screen operand exactly), or, with SKM_FLAG_PRUNE,
+ *        exact dimension pruning over 32-dimension prefix blocks.
  *   SQ8  uint8 [k][d] centroid codes; exact integer code-space distance
  *        sum (xbar_i - cbar_i)^2 (dist is that integer, as float).
  *   RBQ1 float [k][d] decoded centroids; per iteration each centroid is
@@ -197,8 +211,10 @@ int skm_screen_prep(const skm_data *x, void *screen, size_t screen_bytes, void *
  *          ip = (t1 + t2) * fl(1/sqrt d), dist = (nx2 + ny2) - 2 (F ip)
  *        where P = sum_i xbar_i ybar_i is an exact AND+popcount sum.
  *  assign int32[n] (required); dist float[n] (may be NULL).
- *  prev_assign int32[n] or NULL: BF16 only, seeds the pruning bound with
- *  the distance to the previous centroid (results do not depend on it).
+ *  prev_assign int32[n] or NULL: with SKM_FLAG_PRUNE, seeds each row's
+ *  pruning bound with the distance to its previous centroid (entries outside
+ *  [0, k) seed with centroid 0; results do not depend on it).  May alias
+ *  `assign`.
  * ------------------------------------------------------------------------ */
 int skm_assign(const skm_data *x, const void *C, int k, const int32_t *prev_assign,
                int32_t *assign, float *dist, void *ws, size_t ws_bytes, void *stream);

@@ -21,6 +21,7 @@ __all__ = [
 ]
 
 REPR_F32, REPR_SQ8, REPR_RBQ1, REPR_BF16 = 0, 1, 2, 3
+FLAG_PRUNE = 1
 DTYPE_F32, DTYPE_BF16 = 0, 1
 OP_ASSIGN, OP_UPDATE, OP_FIT, OP_QUANTIZE, OP_PCA = 0, 1, 2, 3, 4
 
@@ -51,7 +52,7 @@ class Data(ctypes.Structure):
         ("repr", ctypes.c_int32), ("d", ctypes.c_int32), ("n", ctypes.c_int64),
         ("x", ctypes.c_void_p), ("nx2", ctypes.c_void_p), ("F", ctypes.c_void_p),
         ("popx", ctypes.c_void_p), ("m", ctypes.c_void_p), ("rbq1_exp", ctypes.c_int32),
-        ("reserved0", ctypes.c_int32), ("screen", ctypes.c_void_p),
+        ("flags", ctypes.c_int32), ("screen", ctypes.c_void_p),
     ]
 
 
@@ -65,7 +66,8 @@ class QuantParams(ctypes.Structure):
 
 class Stats(ctypes.Structure):
     _fields_ = [("rescored_rows", ctypes.c_int64), ("fallback_rows", ctypes.c_int64),
-                ("empty_clusters", ctypes.c_int64), ("reserved", ctypes.c_int64 * 5)]
+                ("empty_clusters", ctypes.c_int64), ("prune_first_block", ctypes.c_int64),
+                ("prune_complete", ctypes.c_int64), ("reserved", ctypes.c_int64 * 3)]
 
 
 class FitConfig(ctypes.Structure):
@@ -140,15 +142,20 @@ def _dev(t):
 class Points:
     """Keeps the tensors of one skm_data alive; `.ref` is the ctypes struct."""
 
-    def __init__(self, repr_, x, d, nx2=None, F=None, popx=None, m=None, rbq1_exp=0, screen=None):
+    def __init__(self, repr_, x, d, nx2=None, F=None, popx=None, m=None, rbq1_exp=0, screen=None, flags=0):
         assert x.is_contiguous()
         self.repr, self.x, self.d = repr_, x, int(d)
         self.nx2, self.F, self.popx, self.m = nx2, F, popx, m
         self.n = x.shape[0]
         self.rbq1_exp = int(rbq1_exp)
         self.screen = screen
+        self.flags = int(flags)
         self.ref = Data(repr_, self.d, self.n, x.data_ptr(), _ptr(nx2), _ptr(F), _ptr(popx), _ptr(m),
-                        self.rbq1_exp, 0, _ptr(screen))
+                        self.rbq1_exp, self.flags, _ptr(screen))
+
+    def with_flags(self, flags):
+        return Points(self.repr, self.x, self.d, self.nx2, self.F, self.popx, self.m, self.rbq1_exp, self.screen,
+                      flags)
 
     def with_screen(self, stream=None):
         """Builds the screening copy once (skm_screen_prep) and attaches it."""
@@ -157,7 +164,8 @@ class Points:
             return self
         buf = _ws(nbytes, self.device)
         _check(lib().skm_screen_prep(ctypes.byref(self.ref), _ptr(buf), buf.numel(), _stream(stream)))
-        return Points(self.repr, self.x, self.d, self.nx2, self.F, self.popx, self.m, self.rbq1_exp, buf)
+        return Points(self.repr, self.x, self.d, self.nx2, self.F, self.popx, self.m, self.rbq1_exp, buf,
+                      self.flags)
 
     @property
     def device(self):
@@ -318,7 +326,8 @@ def skm_fit(pts: Points, k, iters, C_init=None, init_idx=None, want_objective=Tr
     _check(lib().skm_fit(ctypes.byref(cfg), ctypes.byref(pts.ref), _ptr(C_init), _ptr(init_idx), _ptr(C),
                          _ptr(assign), _ptr(dist), obj, ctypes.byref(st), _ptr(ws), ws.numel(), _stream(stream)))
     stats = {"rescored_rows": st.rescored_rows, "fallback_rows": st.fallback_rows,
-             "empty_clusters": st.empty_clusters}
+             "empty_clusters": st.empty_clusters, "prune_first_block": st.prune_first_block,
+             "prune_complete": st.prune_complete}
     return C, assign, dist, (list(obj) if obj is not None else None), stats
 
 

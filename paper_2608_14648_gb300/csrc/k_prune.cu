@@ -1,0 +1,182 @@
+// Exact dimension pruning (Section 3.1 "SuperKMeans": partial distances over
+// prefix blocks of the projected dimensions; a centroid is dropped once its
+// partial distance exceeds the row's current best).  CUDA cores, fp32.
+//
+// One warp per point row.  The bound beta starts at the exact distance to a
+// seed centroid (the previous assignment when given, else centroid 0).
+// Centroids are taken 256 at a time: lane l computes the first 32-dimension
+// block of centroid c0 + 32 s + l, the survivors (partial <= beta * slack) are
+// compacted into a shared-memory queue with __ballot_sync / __popc, and each
+// further block re-filters the queue the same way.  Candidates that complete
+// all blocks carry their full distance; the warp keeps the smallest (ties to
+// the lowest index).  Partial sums only grow block by block and every term is
+// non-negative, so dropping a centroid whose partial already exceeds beta
+// never drops the nearest one; `slack` covers the fp32 rounding of the sums,
+// so the result is the exact fp32 argmin whatever the seed.
+#include "skm_internal.cuh"
+
+namespace skm {
+namespace {
+
+constexpr int PR_WARPS = 4;  // 32 KiB of static shared memory per block
+constexpr int PR_BATCH = 256;
+constexpr int PR_MAX_D = 1024;
+
+template <typename TX>
+__device__ __forceinline__ float ldx(const TX *p);
+template <>
+__device__ __forceinline__ float ldx<float>(const float *p) {
+    return __ldg(p);
+}
+template <>
+__device__ __forceinline__ float ldx<uint16_t>(const uint16_t *p) {
+    return __uint_as_float(((uint32_t)__ldg(p)) << 16);
+}
+
+// sum over dims [32b, min(32b + 32, d)) of (x_i - c_i)^2, in increasing i
+__device__ __forceinline__ float block_partial(const float *sx, const float *c, int d, int b) {
+    float s = 0.0f;
+    const int i0 = 32 * b;
+    if (i0 + 32 <= d && (d % 4) == 0) {
+        const float4 *c4 = reinterpret_cast<const float4 *>(c + i0);
+#pragma unroll
+        for (int q = 0; q < 8; ++q) {
+            const float4 cv = __ldg(c4 + q);
+            float t = __fsub_rn(sx[i0 + 4 * q], cv.x);
+            s = __fmaf_rn(t, t, s);
+            t = __fsub_rn(sx[i0 + 4 * q + 1], cv.y);
+            s = __fmaf_rn(t, t, s);
+            t = __fsub_rn(sx[i0 + 4 * q + 2], cv.z);
+            s = __fmaf_rn(t, t, s);
+            t = __fsub_rn(sx[i0 + 4 * q + 3], cv.w);
+            s = __fmaf_rn(t, t, s);
+        }
+    } else {
+        const int i1 = min(d, i0 + 32);
+        for (int i = i0; i < i1; ++i) {
+            const float t = __fsub_rn(sx[i], __ldg(c + i));
+            s = __fmaf_rn(t, t, s);
+        }
+    }
+    return s;
+}
+
+template <typename TX>
+__global__ void __launch_bounds__(PR_WARPS * 32) prune_assign_kernel(
+    const TX *__restrict__ X, int64_t n, int d, const float *__restrict__ C, int k,
+    const int32_t *__restrict__ prev, int32_t *__restrict__ assign, float *__restrict__ dist,
+    unsigned long long *__restrict__ counters) {
+    __shared__ float sx_all[PR_WARPS][PR_MAX_D];
+    __shared__ int qid[PR_WARPS][2][PR_BATCH];
+    __shared__ float qps[PR_WARPS][2][PR_BATCH];
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const unsigned lt = (1u << lane) - 1u;
+    float *sx = sx_all[warp];
+    const int nb = (d + 31) >> 5;
+    // relative rounding of a d-term fp32 sum of non-negative terms is below
+    // d * 2^-24; keep anything within twice that of beta
+    const float slack = 1.0f + 2.0f * (float)(d + 1) * 0x1p-24f;
+    const int64_t nw = (int64_t)gridDim.x * PR_WARPS;
+    unsigned long long first_alive = 0, complete = 0;
+    for (int64_t row = (int64_t)blockIdx.x * PR_WARPS + warp; row < n; row += nw) {
+        __syncwarp();
+        for (int i = lane; i < d; i += 32) sx[i] = ldx<TX>(X + row * d + i);
+        __syncwarp();
+        int best = prev ? prev[row] : 0;
+        if (best < 0 || best >= k) best = 0;
+        float beta = 0.0f;
+        for (int b = 0; b < nb; ++b) beta += block_partial(sx, C + (int64_t)best * d, d, b);
+        for (int c0 = 0; c0 < k; c0 += PR_BATCH) {
+            __syncwarp();  // queue 0 may still be read by the previous batch
+            // first block over the whole batch, survivors compacted into queue 0
+            int cnt = 0;
+            for (int s = 0; s < PR_BATCH / 32; ++s) {
+                const int j = c0 + 32 * s + lane;
+                const float p = (j < k) ? block_partial(sx, C + (int64_t)j * d, d, 0) : INFINITY;
+                const bool alive = p <= beta * slack;
+                const unsigned m = __ballot_sync(0xffffffffu, alive);
+                if (alive) {
+                    const int pos = cnt + __popc(m & lt);
+                    qid[warp][0][pos] = j;
+                    qps[warp][0][pos] = p;
+                }
+                cnt += __popc(m);
+            }
+            first_alive += cnt;
+            int src = 0;
+            for (int b = 1; b < nb && cnt > 0; ++b) {
+                __syncwarp();
+                int ncnt = 0;
+                for (int t0 = 0; t0 < cnt; t0 += 32) {
+                    const int t = t0 + lane;
+                    const bool valid = t < cnt;
+                    const int j = valid ? qid[warp][src][t] : 0;
+                    const float p =
+                        valid ? qps[warp][src][t] + block_partial(sx, C + (int64_t)j * d, d, b) : INFINITY;
+                    const bool alive = valid && p <= beta * slack;
+                    const unsigned m = __ballot_sync(0xffffffffu, alive);
+                    if (alive) {
+                        const int pos = ncnt + __popc(m & lt);
+                        qid[warp][src ^ 1][pos] = j;
+                        qps[warp][src ^ 1][pos] = p;
+                    }
+                    ncnt += __popc(m);
+                }
+                cnt = ncnt;
+                src ^= 1;
+            }
+            __syncwarp();
+            complete += cnt;
+            // complete candidates: full distances; keep the smallest (lowest index on ties)
+            for (int t0 = 0; t0 < cnt; t0 += 32) {
+                const int t = t0 + lane;
+                float p = INFINITY;
+                int j = 0x7fffffff;
+                if (t < cnt) {
+                    p = qps[warp][src][t];
+                    j = qid[warp][src][t];
+                }
+#pragma unroll
+                for (int o = 16; o > 0; o >>= 1) {
+                    const float op = __shfl_xor_sync(0xffffffffu, p, o);
+                    const int oj = __shfl_xor_sync(0xffffffffu, j, o);
+                    if (op < p || (op == p && oj < j)) {
+                        p = op;
+                        j = oj;
+                    }
+                }
+                if (p < beta || (p == beta && j < best)) {
+                    beta = p;
+                    best = j;
+                }
+            }
+        }
+        if (lane == 0) {
+            assign[row] = best;
+            if (dist) dist[row] = beta;
+        }
+    }
+    if (counters && lane == 0) {
+        atomicAdd(&counters[0], first_alive);
+        atomicAdd(&counters[1], complete);
+    }
+}
+
+}  // namespace
+
+cudaError_t launch_prune_assign(const void *X, int x_is_bf16, int64_t n, int d, const float *C,
+                                int k, const int32_t *prev, int32_t *assign, float *dist,
+                                unsigned long long *counters, cudaStream_t st) {
+    if (n == 0) return cudaSuccess;
+    int64_t blocks = (n + PR_WARPS - 1) / PR_WARPS;
+    if (blocks > 152 * 16) blocks = 152 * 16;
+    if (x_is_bf16)
+        prune_assign_kernel<uint16_t><<<(int)blocks, PR_WARPS * 32, 0, st>>>(
+            static_cast<const uint16_t *>(X), n, d, C, k, prev, assign, dist, counters);
+    else
+        prune_assign_kernel<float><<<(int)blocks, PR_WARPS * 32, 0, st>>>(
+            static_cast<const float *>(X), n, d, C, k, prev, assign, dist, counters);
+    return launched();
+}
+
+}  // namespace skm

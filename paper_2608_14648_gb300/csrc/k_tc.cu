@@ -1063,6 +1063,7 @@ void tc_plan(int repr, int64_t n, int d, int k, const void *x, const void *scree
              TcAssignBufs &b) {
     b.stats = cv.take<int64_t>(4);
     b.counters = cv.take<int32_t>(4);
+    if (repr < 0) return;  // statistics only
     const int dp = round8(d);
     const bool dense = repr == SKM_REPR_F32 || repr == SKM_REPR_BF16 ||
                        (repr == SKM_REPR_RBQ1 && d <= TC_RBQ1_MAX_D) ||

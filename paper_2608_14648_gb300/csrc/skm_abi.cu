@@ -36,7 +36,8 @@ constexpr int MAX_D = 4096;
 constexpr int MAX_K = 65536;
 constexpr int64_t MAX_N = (int64_t(1) << 31) - 1;
 constexpr int64_t MAX_N_RBQ1 = int64_t(1) << 24;
-constexpr int RED_BLOCKS = 304;  // 2 x 152 SMs for column / objective reductions
+constexpr int RED_BLOCKS = 304;
+constexpr int PRUNE_MAX_D = 1024;  // 2 x 152 SMs for column / objective reductions
 
 static int check_data(const skm_data *x, bool need_codes = true) {
     if (!x) return set_error(SKM_ERR_INVALID_ARG, "skm_data is NULL");
@@ -49,6 +50,9 @@ static int check_data(const skm_data *x, bool need_codes = true) {
         return set_error(x->n < 1 ? SKM_ERR_INVALID_ARG : SKM_ERR_UNSUPPORTED,
                          "n = %lld outside [1, 2^31)", (long long)x->n);
     if (need_codes && !x->x) return set_error(SKM_ERR_INVALID_ARG, "x->x is NULL");
+    if ((x->flags & SKM_FLAG_PRUNE) && (x->repr == SKM_REPR_F32 || x->repr == SKM_REPR_BF16) &&
+        x->d > PRUNE_MAX_D)
+        return set_error(SKM_ERR_UNSUPPORTED, "SKM_FLAG_PRUNE supports d <= %d", PRUNE_MAX_D);
     if (x->repr == SKM_REPR_RBQ1) {
         if (x->n > MAX_N_RBQ1)
             return set_error(SKM_ERR_UNSUPPORTED, "RBQ1 supports n <= 2^24 (got %lld)",
@@ -69,7 +73,12 @@ static int check_k(const skm_data *x, int k, bool k_le_n = false) {
 }
 
 // ------------------------------------------------------------ workspace plans
+static bool use_prune(const skm_data *x) {
+    return (x->flags & SKM_FLAG_PRUNE) && (x->repr == SKM_REPR_F32 || x->repr == SKM_REPR_BF16);
+}
+
 struct AssignBufs {
+    unsigned long long *prune = nullptr;    // [0] pairs alive after block 1, [1] complete
     int32_t *nx = nullptr, *nc = nullptr;  // SQ8 with d > 1024 (__dp4a path)
     uint4 *planes = nullptr;                // RBQ1 with d > 1024 (AND + popcount path)
     Rbq1CInfo *info = nullptr;
@@ -79,6 +88,11 @@ struct AssignBufs {
 static void plan_assign(const skm_data *x, int k, Carver &cv, AssignBufs &b) {
     const int64_t n = x->n;
     const int d = x->d;
+    b.prune = cv.take<unsigned long long>(2);
+    if (use_prune(x)) {
+        tc_plan(-1, n, d, k, x->x, x->screen, cv, b.tc);  // statistics only
+        return;
+    }
     switch (x->repr) {
     case SKM_REPR_SQ8:
         if (d > TC_SQ8_MAX_D) {
@@ -157,6 +171,12 @@ static int do_assign(const skm_data *x, const void *C, int k, const int32_t *pre
                      int32_t *assign, float *dist, AssignBufs &b, cudaStream_t st) {
     const int64_t n = x->n;
     const int d = x->d;
+    if (use_prune(x)) {
+        SKM_CUDA_TRY(launch_prune_assign(x->x, x->repr == SKM_REPR_BF16, n, d,
+                                         static_cast<const float *>(C), k, prev, assign, dist,
+                                         b.prune, st));
+        return SKM_OK;
+    }
     switch (x->repr) {
     case SKM_REPR_F32:
         SKM_TRY(tc_assign_float(x, static_cast<const float *>(C), k, assign, dist, b.tc, st));
@@ -499,6 +519,7 @@ int skm_fit(const skm_fit_config *cfg, const skm_data *x, const void *C_init,
         xd.screen = b.screen;
     }
     SKM_TRY(tc_init_stats(b.a.tc, st));
+    SKM_CUDA_TRY(cudaMemsetAsync(b.a.prune, 0, 2 * sizeof(unsigned long long), st));
     int e = 0;
     if (x->repr == SKM_REPR_RBQ1) {
         SKM_CUDA_TRY(launch_rbq1_exponent(x->F, n, b.maxbits, b.e_dev, st));
@@ -532,9 +553,8 @@ int skm_fit(const skm_fit_config *cfg, const skm_data *x, const void *C_init,
     int32_t *assign = assign_out;
     for (int it = 0; it <= cfg->iters; ++it) {
         const bool want_obj = objective_host != nullptr;
-        SKM_TRY(do_assign(&xd, C_out, k, nullptr, assign, (want_obj || it == cfg->iters) ? dist
-                                                                                          : nullptr,
-                          b.a, st));
+        SKM_TRY(do_assign(&xd, C_out, k, it > 0 ? assign : nullptr, assign,
+                          (want_obj || it == cfg->iters) ? dist : nullptr, b.a, st));
         if (want_obj) {
             SKM_CUDA_TRY(launch_sum_float_to_double(dist, n, b.partials, nblk, st));
             SKM_CUDA_TRY(launch_sum_double(b.partials, nblk, b.sum, st));
@@ -548,6 +568,10 @@ int skm_fit(const skm_fit_config *cfg, const skm_data *x, const void *C_init,
     skm_stats local;
     memset(&local, 0, sizeof(local));
     SKM_TRY(tc_read_stats(b.a.tc, &local, st));
+    unsigned long long pr[2] = {0, 0};
+    SKM_CUDA_TRY(cudaMemcpy(pr, b.a.prune, sizeof(pr), cudaMemcpyDeviceToHost));
+    local.prune_first_block = (int64_t)pr[0];
+    local.prune_complete = (int64_t)pr[1];
     if (stats_host) {
         *stats_host = local;
         std::vector<int64_t> cnt(k);

@@ -316,3 +316,51 @@ def test_sharded_update_matches_single(skm, repr_name):
         assert float(rel.max()) <= 1e-5
     else:
         assert torch.equal(C_merged, C_single)
+
+
+# -------------------------------------------------- exact dimension pruning
+@pytest.mark.parametrize("repr_name,n,d,k", [("bf16", 3000, 256, 300), ("bf16", 777, 64, 13),
+                                             ("f32", 2000, 768, 200), ("f32", 500, 33, 40)])
+def test_prune_assign_vs_oracle_and_seed_independent(skm, repr_name, n, d, k):
+    X = _points(n, d, seed=n + k)
+    if repr_name == "bf16":
+        Xd = X.to(DEV).to(torch.bfloat16).view(torch.int16)
+        xb = Xd.cpu().numpy().view(np.uint16)
+        C = oracle.bf16_to_f32(xb[synth.forgy_indices(n, k, seed=4).numpy()]).copy()
+        pts = skm.Points(skm.REPR_BF16, Xd, d)
+        a_or, best, second = oracle.assign_bf16(xb, C)
+    else:
+        Xd = X.to(DEV)
+        C = X[synth.forgy_indices(n, k, seed=4)].numpy().copy()
+        pts = skm.Points(skm.REPR_F32, Xd, d)
+        a_or, best, second = oracle.assign_f32(X.numpy(), C)
+    Cd = torch.from_numpy(C).to(DEV)
+    pp = pts.with_flags(skm.FLAG_PRUNE)
+    a0, d0 = skm.skm_assign(pp, Cd)
+    _check_f32(a0.cpu().numpy(), d0.cpu().numpy(), best, second, a_or, f"prune {repr_name}")
+    # the seed of the bound changes the work, never the result
+    prev = torch.randint(0, k, (n,), generator=torch.Generator().manual_seed(7), dtype=torch.int32).to(DEV)
+    a1, d1 = skm.skm_assign(pp, Cd, prev_assign=prev)
+    a2, d2 = skm.skm_assign(pp, Cd, prev_assign=a0.clone())
+    assert torch.equal(a1, a0) and torch.equal(a2, a0)
+    assert torch.equal(d1, d0) and torch.equal(d2, d0)
+    # and the tensor-core screen reaches the same assignment
+    a3, _ = skm.skm_assign(pts, Cd)
+    assert (a3 == a0).float().mean().item() >= AGREE
+
+
+def test_prune_fit_bf16(skm):
+    n, d, k, iters = 6000, 256, 64, 5
+    X = _points(n, d, seed=33)
+    Xd = X.to(DEV).to(torch.bfloat16).view(torch.int16)
+    xb = Xd.cpu().numpy().view(np.uint16)
+    idx = synth.forgy_indices(n, k, seed=33)
+    C0 = oracle.bf16_to_f32(xb[idx.numpy()]).copy()
+    pts = skm.Points(skm.REPR_BF16, Xd, d, flags=skm.FLAG_PRUNE)
+    C, a, _, obj, stats = skm.skm_fit(pts, k, iters, C_init=torch.from_numpy(C0).to(DEV))
+    Co, ao, objo = oracle.lloyd_bf16(xb, C0, iters)
+    assert (a.cpu().numpy() == ao).mean() >= AGREE
+    assert abs(obj[-1] - objo[-1]) / objo[-1] <= 1e-4
+    total = n * k * (iters + 1)
+    print("prune stats", stats, "first-block survival", stats["prune_first_block"] / total)
+    assert 0 < stats["prune_complete"] <= stats["prune_first_block"] <= total
