@@ -148,6 +148,8 @@ def run_ours(args):
     if world > 1:
         import torch.distributed as dist
 
+        from paper_2608_14648_gb300 import dist as skd
+
         dist.init_process_group("nccl")
     peaks = load_peaks()
 
@@ -160,14 +162,11 @@ def run_ours(args):
     pts32 = skm.Points(skm.REPR_F32, X, DIM).with_screen()  # bf16 screening copy, built once
     q = skm.skm_quantize(skm.REPR_RBQ1, X)
     if world > 1:  # global mean, then re-encode; global fixed-point exponent
-        dist.all_reduce(q["m"])
-        q["m"] /= world
-        q = skm.skm_quantize(skm.REPR_RBQ1, X, fit=False, m=q["m"])
+        m = skd.global_mean(q["m"].double() * N_POINTS, N_POINTS)
+        q = skm.skm_quantize(skm.REPR_RBQ1, X, fit=False, m=m.contiguous())
     e = skm.skm_rbq1_exponent(q["F"])
     if world > 1:
-        et = torch.tensor([e], device=dev)
-        dist.all_reduce(et, op=dist.ReduceOp.MIN)
-        e = int(et.item())
+        e = skd.global_exponent(e, dev)
     ptsR = skm.rbq1_points(q, DIM, e).with_screen()  # e4m3 expansion of the bits, built once
     Cr, _, _, _, _ = skm.skm_fit(ptsR, K, 0, init_idx=idx, want_objective=False, want_dist=False)
     if world > 1:
@@ -200,8 +199,7 @@ def run_ours(args):
             part.zero_()
             cnt.zero_()
             skm.skm_update(pts, a, None, counts=cnt, partial=part, ws=wsU)
-            dist.all_reduce(part)
-            dist.all_reduce(cnt)
+            skd.allreduce_partials(part, cnt)
             skm.skm_update_finalize(pts, part, cnt, C)
 
     def step(record):

@@ -1,0 +1,221 @@
+"""Parity at the full workload sizes, through the C ABI, in the launch
+configuration bench.py uses (screening copies built once, skm_assign /
+skm_update per iteration).  Outputs are checked on sampled rows the oracle
+computes one by one (bit-exact for integer paths), updates on all rows or on
+whole clusters, objectives in full where the oracle affords it."""
+import math
+
+import numpy as np
+import pytest
+import torch
+
+import oracle
+import synth
+
+pytestmark = pytest.mark.gpu
+DEV = "cuda"
+AGREE, GAP_TOL = 0.999, 1e-5
+
+
+@pytest.fixture(scope="module")
+def skm(cuda_ok):
+    import paper_2608_14648_gb300 as skm
+
+    skm.lib()
+    return skm
+
+
+def _sample(n, m, seed):
+    return np.sort(np.random.default_rng(seed).choice(n, size=m, replace=False))
+
+
+def _check_float(a_gpu, d_gpu, a_or, best, second, what):
+    agree = a_gpu == a_or
+    assert agree.mean() >= AGREE, f"{what}: agreement {agree.mean()}"
+    if not agree.all():
+        gap = (second - best) / np.maximum(best, 1e-30)
+        assert np.all(gap[~agree] <= GAP_TOL), f"{what}: gap {gap[~agree].max()}"
+    if d_gpu is not None:
+        np.testing.assert_allclose(d_gpu[agree], best[agree], rtol=2e-5, atol=1e-6)
+
+
+def _cluster_subset_update(codes_or_x, assign, clusters):
+    """Rows of the given clusters, with assignments renumbered 0..len-1."""
+    sel = np.isin(assign, clusters)
+    remap = {c: i for i, c in enumerate(clusters)}
+    return codes_or_x[sel], np.array([remap[a] for a in assign[sel]], np.int32)
+
+
+def test_emb1m_d768_f32_and_rbq1(skm):
+    spec = synth.WORKLOADS["emb1m_d768"]
+    n, d, k = spec.n, spec.d, spec.k
+    X = synth.workload_points(spec, seed=0, device=DEV)
+    idx = synth.forgy_indices(n, k, seed=0).to(DEV)
+    C = X[idx].clone()
+    rows = _sample(n, 2000, 1)
+    Xs = X[torch.from_numpy(rows).to(DEV)].cpu().numpy()
+
+    # fp32: two Lloyd iterations, then parity of the third assignment
+    pts = skm.Points(skm.REPR_F32, X, d).with_screen()
+    for _ in range(2):
+        a, _ = skm.skm_assign(pts, C, want_dist=False)
+        skm.skm_update(pts, a, C)
+    a, dist = skm.skm_assign(pts, C)
+    Ch = C.cpu().numpy()
+    a_or, best, second = oracle.assign_f32(Xs, Ch)
+    _check_float(a.cpu().numpy()[rows], dist.cpu().numpy()[rows], a_or, best, second, "emb1m f32")
+    # update with identical assignments, all rows
+    Xh = X.cpu().numpy()
+    ah = a.cpu().numpy()
+    Cn, counts = skm.skm_update(pts, a, C.clone())
+    Co, co = oracle.update_f32(Xh, ah, Ch)
+    np.testing.assert_array_equal(counts.cpu().numpy(), co)
+    rel = np.linalg.norm(Cn.cpu().numpy() - Co, axis=1) / np.maximum(np.linalg.norm(Co, axis=1), 1e-30)
+    assert rel.max() <= 1e-4
+    obj = skm.skm_objective(X, C, a)
+    objo = oracle.objective_f32(Xh, Ch, ah)
+    assert abs(obj - objo) / objo <= 1e-4
+
+    # 1-bit: encode, one iteration, assignment and update bit-exact
+    q = skm.skm_quantize(skm.REPR_RBQ1, X)
+    ptsR = skm.rbq1_points(q, d).with_screen()
+    h = {kk: v.cpu().numpy() for kk, v in q.items()}
+    codes = h["codes"].view(np.uint32)
+    c2, nx2, F, popx = oracle.rbq1_encode(Xs, h["m"])
+    np.testing.assert_array_equal(codes[rows], c2)
+    np.testing.assert_allclose(h["F"][rows], F, rtol=1e-6)
+    Cr = C.clone()
+    aR, estR = skm.skm_assign(ptsR, Cr)
+    prep = oracle.rbq1_centroid_sq4(Cr.cpu().numpy(), h["m"])
+    ao, esto = oracle.rbq1_assign(codes[rows], h["nx2"][rows], h["F"][rows], h["popx"][rows], d, prep)
+    np.testing.assert_array_equal(aR.cpu().numpy()[rows], ao)
+    np.testing.assert_array_equal(estR.cpu().numpy()[rows], esto)
+    CrN, cntR = skm.skm_update(ptsR, aR, Cr.clone())
+    CroN, cro = oracle.rbq1_update(codes, h["F"], d, h["m"], ptsR.rbq1_exp, aR.cpu().numpy(), Cr.cpu().numpy())
+    np.testing.assert_array_equal(cntR.cpu().numpy(), cro)
+    np.testing.assert_array_equal(CrN.cpu().numpy(), CroN)
+    del X, pts, ptsR
+    torch.cuda.empty_cache()
+
+
+def test_emb1m_d1024_sq8(skm):
+    spec = synth.WORKLOADS["emb1m_d1024_sq8"]
+    n, d, k = spec.n, spec.d, spec.k
+    X = synth.workload_points(spec, seed=0, device=DEV)
+    q = skm.skm_quantize(skm.REPR_SQ8, X)
+    rows = _sample(n, 2000, 2)
+    Xh = X.cpu().numpy()
+    b, s = oracle.sq8_fit(Xh)
+    np.testing.assert_array_equal(q["b"].cpu().numpy(), b)
+    np.testing.assert_array_equal(q["s"].cpu().numpy(), s)
+    codes = q["codes"].cpu().numpy()
+    np.testing.assert_array_equal(codes[rows], oracle.sq8_encode(Xh[rows], b, s))
+    pts = skm.Points(skm.REPR_SQ8, q["codes"], d).with_screen()
+    idx = synth.forgy_indices(n, k, seed=0)
+    Cc = q["codes"][idx.to(DEV)].clone()
+    a, dist = skm.skm_assign(pts, Cc)
+    ao, bo = oracle.assign_sq8(codes[rows], Cc.cpu().numpy())
+    np.testing.assert_array_equal(a.cpu().numpy()[rows], ao)
+    np.testing.assert_array_equal(dist.cpu().numpy()[rows], bo.astype(np.float32))
+    Cn, counts = skm.skm_update(pts, a, Cc.clone())
+    Co, co = oracle.update_sq8(codes, a.cpu().numpy(), Cc.cpu().numpy())
+    np.testing.assert_array_equal(counts.cpu().numpy(), co)
+    np.testing.assert_array_equal(Cn.cpu().numpy(), Co)
+    # SSE in full precision: decoded centroids against the fp32 points
+    Cdec = skm.skm_sq8_decode(Cn, q["b"], q["s"])
+    a2, _ = skm.skm_assign(pts, Cn, want_dist=False)
+    sse = skm.skm_objective(X, Cdec, a2)
+    sseo = oracle.objective_f32(Xh, oracle.sq8_decode(Co, b, s), a2.cpu().numpy())
+    assert abs(sse - sseo) / sseo <= 1e-4
+    del X, pts
+    torch.cuda.empty_cache()
+
+
+def test_emb10m_d1024_rotation_rbq1(skm):
+    spec = synth.WORKLOADS["emb10m_d1024_rbq1"]
+    n, d, k = spec.n, spec.d, spec.k
+    X = synth.workload_points(spec, seed=0, device=DEV)
+    P = synth.haar_rotation(d, 99).to(torch.float32).contiguous()
+    Y = skm.skm_project(X, P.to(DEV))  # the seeded random rotation before 1-bit encoding
+    rows = _sample(n, 500, 3)
+    rt = torch.from_numpy(rows).to(DEV)
+    Yo = oracle.project(X[rt].cpu().numpy(), P.numpy())
+    assert np.max(np.abs(Y[rt].cpu().numpy() - Yo)) < 2e-6
+    del X
+    torch.cuda.empty_cache()
+    q = skm.skm_quantize(skm.REPR_RBQ1, Y)
+    pts = skm.rbq1_points(q, d).with_screen()
+    idx = synth.forgy_indices(n, k, seed=0).to(DEV)
+    C, _, _, _, _ = skm.skm_fit(pts, k, 0, init_idx=idx, want_objective=False, want_dist=False)
+    a, est = skm.skm_assign(pts, C)
+    m = q["m"].cpu().numpy()
+    codes_s = q["codes"][rt].cpu().numpy().view(np.uint32)
+    c2, nx2, F, popx = oracle.rbq1_encode(Y[rt].cpu().numpy(), m)
+    np.testing.assert_array_equal(codes_s, c2)
+    prep = oracle.rbq1_centroid_sq4(C.cpu().numpy(), m)
+    ao, esto = oracle.rbq1_assign(codes_s, q["nx2"][rt].cpu().numpy(), q["F"][rt].cpu().numpy(),
+                                  q["popx"][rt].cpu().numpy(), d, prep)
+    np.testing.assert_array_equal(a[rt].cpu().numpy(), ao)
+    np.testing.assert_array_equal(est[rt].cpu().numpy(), esto)
+    # update: whole clusters 0..7 recomputed by the oracle
+    Cn, counts = skm.skm_update(pts, a, C.clone())
+    ah = a.cpu().numpy()
+    clusters = np.arange(8)
+    sel = np.isin(ah, clusters)
+    codes_all = q["codes"].cpu().numpy().view(np.uint32)
+    Fh = q["F"].cpu().numpy()
+    sub_a = ah[sel].astype(np.int32)
+    Co, co = oracle.rbq1_update(codes_all[sel], Fh[sel], d, m, pts.rbq1_exp, sub_a, C.cpu().numpy()[:8])
+    np.testing.assert_array_equal(counts.cpu().numpy()[:8], co)
+    np.testing.assert_array_equal(Cn.cpu().numpy()[:8], Co)
+    assert int(counts.sum()) == n
+    del Y, pts
+    torch.cuda.empty_cache()
+
+
+def test_emb10m_pca256_bf16(skm):
+    spec = synth.WORKLOADS["emb10m_pca256"]
+    n, D, k, dp = spec.n, spec.d, spec.k, 256
+    X = synth.workload_points(spec, seed=0, device=DEV)
+    mean, P, w = skm.skm_pca_fit(X, dp)
+    Pn = P.double().cpu().numpy()
+    np.testing.assert_allclose(Pn.T @ Pn, np.eye(dp), atol=2e-5)
+    wn = w.cpu().numpy()
+    assert np.all(np.diff(wn) <= 1e-7 * wn[0])
+    # eigenvalues agree with the Rayleigh quotients of an independent subsample
+    sub = X[torch.from_numpy(_sample(n, 100_000, 4)).to(DEV)].cpu().numpy()
+    mu, cov = oracle.mean_cov(sub)
+    rq = np.einsum("ij,ik,kj->j", Pn, cov, Pn)
+    np.testing.assert_allclose(rq, wn, rtol=0.05)
+    Yb = skm.skm_project(X, P, mean, out_dtype=skm.DTYPE_BF16).view(torch.int16)
+    rows = _sample(n, 200, 5)
+    rt = torch.from_numpy(rows).to(DEV)
+    Yo = oracle.project(X[rt].cpu().numpy(), P.cpu().numpy(), mean.cpu().numpy())
+    yb = Yb[rt].cpu().numpy().view(np.uint16)
+    err = np.abs(oracle.bf16_to_f32(yb).astype(np.float64) - Yo)
+    assert np.all(err <= 2.0 ** -8 * np.abs(Yo) + 1e-5)
+    del X
+    torch.cuda.empty_cache()
+    pts = skm.Points(skm.REPR_BF16, Yb, dp).with_screen()
+    idx = synth.forgy_indices(n, k, seed=0).to(DEV)
+    C = (Yb[idx].to(torch.int32) << 16).view(torch.float32).contiguous()
+    a, dist = skm.skm_assign(pts, C)
+    yb_s = Yb[rt].cpu().numpy().view(np.uint16)
+    a_or, best, second = oracle.assign_bf16(yb_s, C.cpu().numpy())
+    _check_float(a[rt].cpu().numpy(), dist[rt].cpu().numpy(), a_or, best, second, "pca256 bf16")
+    # exact pruning gives the same assignment on the sampled rows
+    rows_p = torch.arange(0, 200_000, device=DEV)
+    sub_pts = skm.Points(skm.REPR_BF16, Yb[rows_p].contiguous(), dp, flags=skm.FLAG_PRUNE)
+    ap, _ = skm.skm_assign(sub_pts, C, prev_assign=a[rows_p].contiguous())
+    assert (ap == a[rows_p]).float().mean().item() >= AGREE
+    # update: whole clusters 0..7
+    Cn, counts = skm.skm_update(pts, a, C.clone())
+    ah = a.cpu().numpy()
+    sel = np.isin(ah, np.arange(8))
+    Co, co = oracle.update_bf16(Yb.cpu().numpy().view(np.uint16)[sel], ah[sel].astype(np.int32),
+                                C.cpu().numpy()[:8])
+    np.testing.assert_array_equal(counts.cpu().numpy()[:8], co)
+    rel = np.linalg.norm(Cn.cpu().numpy()[:8] - Co, axis=1) / np.linalg.norm(Co, axis=1)
+    assert rel.max() <= 1e-4
+    del Yb, pts
+    torch.cuda.empty_cache()
