@@ -33,8 +33,16 @@ N_POINTS, DIM, K, N_COMP = 1_000_000, 768, 1000, 2000
 METRIC = "k-means point·centroid distances/s per Lloyd iter (1 GB300); % of roofline"
 WORKLOAD = "emb1m_d768: N=1,000,000 x d=768 unit-norm GMM embeddings, k=1,000; fp32 + RabitQ 1-bit"
 SM_COUNT = 152
-# POPC results per clock per SM used for the 1-bit kernel's ALU roofline.
+# POPC results per clock per SM used for the 1-bit kernel's ALU roofline
+# (measured 15.9 on GB300 with a throughput probe).
 POPC_PER_CLK_SM = 16
+# DRAM bytes (read + write) per point of the assignment kernels, from one ncu
+# capture each (200,000 points x d=768, k=1000; profiles/tc_assign_*.md).
+# Each point row is read once per launch, so traffic scales with the points.
+TRAFFIC_PER_POINT = {
+    "assign_f32": (311.908352e6 + 5.505024e6) / 200_000,
+    "assign_rbq1": (156.861952e6 + 3.515392e6) / 200_000,
+}
 
 
 def env_rank():
@@ -273,8 +281,10 @@ def run_ours(args):
         kd["frac"] = kd["achieved"] / kd["peak"]
     dom = max((n for n in kernels if kernels[n].get("in_step", True)), key=lambda n: kernels[n]["ms"])
     kd = kernels[dom]
+    traffic = TRAFFIC_PER_POINT.get(dom)
     roofline = {"bound": kd["bound"], "achieved": round(kd["achieved"], 4), "peak": round(kd["peak"], 4),
-                "unit": kd["unit"], "frac": round(kd["frac"], 5), "traffic": None, "kernel": dom,
+                "unit": kd["unit"], "frac": round(kd["frac"], 5),
+                "traffic": round(traffic * N_POINTS) if traffic else None, "kernel": dom,
                 "peak_source": f"{peaks['source']} ({'sustained' if long_region else 'burst'} bf16"
                                f"{', x2 for e4m3' if dom == 'assign_rbq1' else ''})"}
 

@@ -205,11 +205,15 @@ int skm_screen_prep(const skm_data *x, void *screen, size_t screen_bytes, void *
  *        sum (xbar_i - cbar_i)^2 (dist is that integer, as float).
  *   RBQ1 float [k][d] decoded centroids; per iteration each centroid is
  *        re-encoded with per-centroid SQ4 (b = min, s = (max-b)/15 of
- *        c - m) and the distance is the estimator of Eq. rabitq_l2 with
+ *        c - m; ny2 = ||c - m||^2 in fp64, pairwise inside 32-dimension
+ *        blocks, blocks added in order) and the distance is the estimator
+ *        of Eq. rabitq_l2 with
  *        Eq. final:rabitq, evaluated in fp32 in the order
- *          t1 = s (2P - sum ybar), t2 = b (2 popx - d),
- *          ip = (t1 + t2) * fl(1/sqrt d), dist = (nx2 + ny2) - 2 (F ip)
- *        where P = sum_i xbar_i ybar_i is an exact AND+popcount sum.
+ *          sd = s fl(1/sqrt d), bd = b fl(1/sqrt d)      (per centroid)
+ *          u = fma(sd, 2P - sum ybar, bd (2 popx - d))
+ *          dist = fma(-2 F, u, nx2 + ny2)
+ *        where P = sum_i xbar_i ybar_i is an exact integer (tensor cores in
+ *        e4m3 for d <= 1024, AND + popcount beyond).
  *  assign int32[n] (required); dist float[n] (may be NULL).
  *  prev_assign int32[n] or NULL: with SKM_FLAG_PRUNE, seeds each row's
  *  pruning bound with the distance to its previous centroid (entries outside

@@ -80,6 +80,7 @@ def lib():
                 "or_project": ([vp, i64, i32, vp, vp, i32, vp], None),
                 "or_mean_cov": ([vp, i64, i32, vp, vp], None),
                 "or_round_bf16": ([vp, i64, vp], None),
+                "or_sumsq_blocked": ([vp, i32], f64),
             }
             for name, (args, res) in sig.items():
                 fn = getattr(L, name)
@@ -258,6 +259,12 @@ def rbq1_centroid_sq4(C, m):
     ny2 = np.empty(k, np.float32)
     lib().or_rbq1_centroid_sq4(_p(C), k, d, _p(_c(m, np.float32)), _p(ybar), _p(b), _p(s), _p(sumy), _p(ny2))
     return ybar, b, s, sumy, ny2
+
+
+def sumsq_blocked(r) -> float:
+    """||r||^2 in the library's blocked fp64 order (see skm_oracle.c)."""
+    r = _c(r, np.float32)
+    return float(lib().or_sumsq_blocked(_p(r), r.size))
 
 
 def rbq1_assign(codes, nx2, F, popx, d, prep):

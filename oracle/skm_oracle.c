@@ -335,22 +335,46 @@ void or_rbq1_encode(const float *X, int64_t n, int d, const float *m, uint32_t *
     }
 }
 
+/* ||rho||^2 in fp64 in a fixed order: per 32-dimension block (zero-padded)
+ * the squares are summed pairwise, v[l] += v[l + o] for o = 16, 8, 4, 2, 1,
+ * and the block sums are added in increasing block order.  The paper fixes
+ * no summation order; this one is the library's, so both sides agree bit for
+ * bit.  Pinned against the sequential fp64 sum (relative 1e-14). */
+static double sumsq_blocked(const float *r, int d) {
+    double q2 = 0.0;
+    for (int w = 0; w < (d + 31) / 32; ++w) {
+        double v[32];
+        for (int l = 0; l < 32; ++l) {
+            int i = 32 * w + l;
+            v[l] = (i < d) ? (double)r[i] * (double)r[i] : 0.0;
+        }
+        for (int o = 16; o >= 1; o >>= 1)
+            for (int l = 0; l < o; ++l) v[l] = v[l] + v[l + o];
+        q2 = q2 + v[0];
+    }
+    return q2;
+}
+
+double or_sumsq_blocked(const float *r, int d) { return sumsq_blocked(r, d); }
+
 /* Centroid side, once per iteration: rho = c - m (fp32); per-centroid SQ4
  * with b = min rho, s = (max rho - b) / 15 (s = 1 when flat); ybar_i =
  * clip(round((rho_i - b) / s), 0, 15) with rounding half to even;
- * sumy = sum ybar; ny2 = ||rho||^2 (fp64, sequential, rounded to fp32). */
+ * sumy = sum ybar; ny2 = ||rho||^2 (fp64, blocked order above, rounded to
+ * fp32). */
 void or_rbq1_centroid_sq4(const float *C, int k, int d, const float *m, uint8_t *ybar,
                           float *b, float *s, int32_t *sumy, float *ny2) {
+    float *rho = (float *)malloc(sizeof(float) * (size_t)d);
     for (int j = 0; j < k; ++j) {
         const float *c = C + (int64_t)j * d;
         float lo = INFINITY, hi = -INFINITY;
-        double q2 = 0.0;
         for (int i = 0; i < d; ++i) {
             float r = c[i] - m[i];
+            rho[i] = r;
             if (r < lo) lo = r;
             if (r > hi) hi = r;
-            q2 += (double)r * (double)r;
         }
+        double q2 = sumsq_blocked(rho, d);
         float sc = (hi - lo) / 15.0f;
         if (!(sc > 0.0f)) sc = 1.0f;
         int32_t sy = 0;
@@ -367,14 +391,16 @@ void or_rbq1_centroid_sq4(const float *C, int k, int d, const float *m, uint8_t 
         sumy[j] = sy;
         ny2[j] = (float)q2;
     }
+    free(rho);
 }
 
-/* Eq. final:rabitq into Eq. rabitq_l2, fp32 in this fixed order:
- *   P   = sum_i xbar_i * ybar_i              (exact integer)
- *   t1  = s * (2P - sum ybar)
- *   t2  = b * (2 popx - d)
- *   ip  = (t1 + t2) * (1/sqrt(d))            (1/sqrt(d) rounded once to fp32)
- *   est = (nx2 + ny2) - 2 (F * ip)
+/* Eq. final:rabitq into Eq. rabitq_l2, fp32, in this fixed order (the paper
+ * fixes none; 1/sqrt(d) is folded into the centroid's SQ4 scale and bias):
+ *   P   = sum_i xbar_i * ybar_i                      (exact integer)
+ *   isd = 1/sqrt(d) rounded once to fp32
+ *   sd  = s * isd,  bd = b * isd                     (per centroid)
+ *   u   = fma(sd, 2P - sum ybar, bd * (2 popx - d))  (= <xbar, y_r - m> estimate)
+ *   est = fma(-2 F, u, nx2 + ny2)                    (Eq. rabitq_l2)
  * argmin over est, ties to the lowest index. */
 void or_rbq1_assign(const uint32_t *codes, const float *nx2, const float *F,
                     const int32_t *popx, int64_t n, int d, const uint8_t *ybar,
@@ -385,6 +411,8 @@ void or_rbq1_assign(const uint32_t *codes, const float *nx2, const float *F,
 #pragma omp parallel for schedule(dynamic, 16)
     for (int64_t p = 0; p < n; ++p) {
         const uint32_t *cw = codes + p * (int64_t)W;
+        const float pc = (float)(2 * popx[p] - d);
+        const float f2 = -2.0f * F[p];
         float best = INFINITY;
         int32_t a = -1;
         for (int j = 0; j < k; ++j) {
@@ -392,12 +420,10 @@ void or_rbq1_assign(const uint32_t *codes, const float *nx2, const float *F,
             int32_t P = 0;
             for (int i = 0; i < d; ++i)
                 if ((cw[i / 32] >> (i % 32)) & 1u) P += y[i];
-            float t1 = s[j] * (float)(2 * P - sumy[j]);
-            float t2 = b[j] * (float)(2 * popx[p] - d);
-            float ip = (t1 + t2) * isd;
-            float nn = nx2[p] + ny2[j];
-            float fi = F[p] * ip;
-            float est = nn - 2.0f * fi;
+            const float sd = s[j] * isd;
+            const float bd = b[j] * isd;
+            const float u = fmaf(sd, (float)(2 * P - sumy[j]), bd * pc);
+            const float est = fmaf(f2, u, nx2[p] + ny2[j]);
             if (est < best) {
                 best = est;
                 a = j;

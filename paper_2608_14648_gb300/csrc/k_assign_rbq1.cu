@@ -3,9 +3,9 @@
 // point code against a 4-bit centroid code is computed exactly as
 // P = sum_w sum_j 2^j popc(xbar_w & plane_j,w) with AND + POPC on packed
 // 32-bit words; the distance estimate follows in fp32 in the fixed order
-//   t1 = s (2P - sumy), t2 = b (2 popx - d), ip = (t1 + t2) * fl(1/sqrt d),
-//   est = (nx2 + ny2) - 2 (F ip)
-// and the argmin keeps the lowest index on ties.
+//   u = fma(sd, 2P - sumy, bd (2 popx - d)),  est = fma(-2 F, u, nx2 + ny2)
+// (sd, bd: the centroid's SQ4 scale and bias times fl(1/sqrt d)), and the
+// argmin keeps the lowest index on ties.
 //
 // One thread per point; the point's code words live in shared memory
 // (transposed, conflict-free), centroid bit planes are staged per chunk and
@@ -21,20 +21,16 @@ __device__ __forceinline__ int plane_dot(uint32_t x, uint4 y) {
     return __popc(x & y.x) + 2 * __popc(x & y.y) + 4 * __popc(x & y.z) + 8 * __popc(x & y.w);
 }
 
-__device__ __forceinline__ float rbq1_estimate(int P, const Rbq1CInfo &ci, float nx2, float F,
-                                               int popx, int d, float isd) {
-    const float t1 = __fmul_rn(ci.s, (float)(2 * P - ci.sumy));
-    const float t2 = __fmul_rn(ci.b, (float)(2 * popx - d));
-    const float ip = __fmul_rn(__fadd_rn(t1, t2), isd);
-    const float nn = __fadd_rn(nx2, ci.ny2);
-    const float fi = __fmul_rn(F, ip);
-    return __fsub_rn(nn, __fmul_rn(2.0f, fi));
+__device__ __forceinline__ float rbq1_estimate(int P, const Rbq1CInfo &ci, float nx2, float f2,
+                                               float pc) {
+    const float u = __fmaf_rn(ci.sd, __int2float_rn(2 * P - ci.sumy), __fmul_rn(ci.bd, pc));
+    return __fmaf_rn(f2, u, __fadd_rn(nx2, ci.ny2));
 }
 
 __global__ void __launch_bounds__(RBQ1_THREADS) assign_rbq1_kernel(
     const uint32_t *__restrict__ codes, const float *__restrict__ nx2, const float *__restrict__ F,
     const int32_t *__restrict__ popx, int64_t n, int d, const uint4 *__restrict__ planes,
-    const Rbq1CInfo *__restrict__ info, int k, int kc, float isd, int32_t *__restrict__ assign,
+    const Rbq1CInfo *__restrict__ info, int k, int kc, int32_t *__restrict__ assign,
     float *__restrict__ dist) {
     extern __shared__ __align__(16) unsigned char smem_raw[];
     const int W = (d + 31) >> 5;
@@ -52,8 +48,8 @@ __global__ void __launch_bounds__(RBQ1_THREADS) assign_rbq1_kernel(
         xs[w * RBQ1_THREADS + t] = (q < n) ? codes[q * W + w] : 0u;
     }
     const float my_nx2 = valid ? nx2[p] : 0.0f;
-    const float my_F = valid ? F[p] : 0.0f;
-    const int my_pop = valid ? popx[p] : 0;
+    const float my_f2 = valid ? __fmul_rn(-2.0f, F[p]) : 0.0f;  // exact
+    const float my_pc = valid ? __int2float_rn(2 * popx[p] - d) : 0.0f;
 
     float best = INFINITY;
     int besti = 0;
@@ -77,7 +73,7 @@ __global__ void __launch_bounds__(RBQ1_THREADS) assign_rbq1_kernel(
             const int Ps[4] = {P0, P1, P2, P3};
 #pragma unroll
             for (int q = 0; q < 4; ++q) {
-                const float est = rbq1_estimate(Ps[q], is[j + q], my_nx2, my_F, my_pop, d, isd);
+                const float est = rbq1_estimate(Ps[q], is[j + q], my_nx2, my_f2, my_pc);
                 if (est < best) {
                     best = est;
                     besti = c0 + j + q;
@@ -88,7 +84,7 @@ __global__ void __launch_bounds__(RBQ1_THREADS) assign_rbq1_kernel(
             int P = 0;
             const uint4 *pj = ps + (size_t)j * W;
             for (int w = 0; w < W; ++w) P += plane_dot(xs[w * RBQ1_THREADS + tid], pj[w]);
-            const float est = rbq1_estimate(P, is[j], my_nx2, my_F, my_pop, d, isd);
+            const float est = rbq1_estimate(P, is[j], my_nx2, my_f2, my_pc);
             if (est < best) {
                 best = est;
                 besti = c0 + j;
@@ -117,9 +113,8 @@ cudaError_t launch_assign_rbq1(const uint32_t *codes, const float *nx2, const fl
     cudaError_t e = cudaFuncSetAttribute(assign_rbq1_kernel,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
-    const float isd = (float)(1.0 / sqrt((double)d));
     assign_rbq1_kernel<<<(unsigned)((n + RBQ1_THREADS - 1) / RBQ1_THREADS), RBQ1_THREADS, smem,
-                         st>>>(codes, nx2, F, popx, n, d, planes, info, k, kc, isd, assign, dist);
+                         st>>>(codes, nx2, F, popx, n, d, planes, info, k, kc, assign, dist);
     return launched();
 }
 

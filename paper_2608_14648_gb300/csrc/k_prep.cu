@@ -4,7 +4,7 @@
 //  s = 1 when flat, ybar = clip(rint((rho - b)/s), 0, 15)) and stored as four
 //  bit planes per 32-dimension word, so that sum_i xbar_i ybar_i =
 //  sum_j 2^j popc(xbar & plane_j), and/or as e4m3 bytes for the tensor kernel.
-//  ||rho||^2 is summed in fp64 in increasing dimension order by one lane.
+//  ||rho||^2 is summed in fp64 in the library's blocked pairwise order.
 //  SQ8: per-row sums of squared codes (exact int32).
 #include "skm_internal.cuh"
 
@@ -13,7 +13,8 @@ namespace skm {
 // One warp per centroid.  rho = c - m is kept in the warp's slice of shared
 // memory; min/max and the code sum are exact warp reductions, the codes of
 // 32 consecutive dimensions become four bit planes through __ballot_sync, and
-// one lane forms ||rho||^2 in fp64 in increasing dimension order.
+// ||rho||^2 is summed in fp64 pairwise inside each 32-dimension block (xor
+// butterfly 16, 8, 4, 2, 1) with the block sums added in order.
 constexpr int CPREP_WARPS = 4;
 
 // e4m3 encodings of the integers 0..15 (sign 0, exponent bias 7, 3 mantissa
@@ -30,7 +31,8 @@ __device__ __forceinline__ uint8_t e4m3_of_code(uint32_t y) {
 // kernel).
 __global__ void __launch_bounds__(CPREP_WARPS * 32) rbq1_cprep_kernel(
     const float *__restrict__ C, int k, int d, const float *__restrict__ m,
-    uint4 *__restrict__ planes, Rbq1CInfo *__restrict__ info, uint8_t *__restrict__ yq, int dq) {
+    uint4 *__restrict__ planes, Rbq1CInfo *__restrict__ info, uint8_t *__restrict__ yq, int dq,
+    float isd) {
     extern __shared__ float sh_rho[];  // [CPREP_WARPS][d]
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int j = blockIdx.x * CPREP_WARPS + warp;
@@ -54,8 +56,13 @@ __global__ void __launch_bounds__(CPREP_WARPS * 32) rbq1_cprep_kernel(
     if (!(sc > 0.0f)) sc = 1.0f;
     const int W = (d + 31) >> 5;
     int32_t sy = 0;
+    double q2 = 0.0;  // ||rho||^2: pairwise within 32-dim blocks, blocks in order
     for (int w = 0; w < W; ++w) {
         const int i = 32 * w + lane;
+        double sq = (i < d) ? __dmul_rn((double)rho[i], (double)rho[i]) : 0.0;
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) sq = __dadd_rn(sq, __shfl_xor_sync(0xffffffffu, sq, o));
+        q2 = __dadd_rn(q2, sq);
         uint32_t y = 0;
         if (i < d) {
             float q = rintf(__fdiv_rn(__fsub_rn(rho[i], lo), sc));
@@ -74,11 +81,9 @@ __global__ void __launch_bounds__(CPREP_WARPS * 32) rbq1_cprep_kernel(
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) sy += __shfl_xor_sync(0xffffffffu, sy, o);
     if (lane == 0) {
-        double q2 = 0.0;
-        for (int i = 0; i < d; ++i) q2 = __dadd_rn(q2, __dmul_rn((double)rho[i], (double)rho[i]));
         Rbq1CInfo in;
-        in.b = lo;
-        in.s = sc;
+        in.bd = __fmul_rn(lo, isd);
+        in.sd = __fmul_rn(sc, isd);
         in.sumy = sy;
         in.ny2 = __double2float_rn(q2);
         info[j] = in;
@@ -94,7 +99,7 @@ static cudaError_t launch_cprep_common(const float *C, int k, int d, const float
         if (e != cudaSuccess) return e;
     }
     rbq1_cprep_kernel<<<(k + CPREP_WARPS - 1) / CPREP_WARPS, CPREP_WARPS * 32, smem, st>>>(
-        C, k, d, m, planes, info, yq, dq);
+        C, k, d, m, planes, info, yq, dq, rbq1_isd(d));
     return launched();
 }
 

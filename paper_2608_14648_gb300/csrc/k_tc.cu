@@ -75,13 +75,12 @@ struct TcParams {
     const int32_t *nx;  // SQ8: centred ||x||^2
     const int32_t *nc;  // SQ8: centred ||c||^2, padded to 256 with a large value
     float *dist;        // SQ8 / RBQ1 (may be null)
-    const float4 *rinfo;     // RBQ1: per column pair (b x2, s x2), padded
+    const float4 *rinfo;     // RBQ1: per column pair (bd x2, sd x2), padded
     const float4 *rinfoq;    // RBQ1: per column pair (-sum ybar x2, ||c - m||^2 x2)
     const float *nx2;        // RBQ1 per point
     const float *F;
     const int32_t *popx;
     int d;
-    float isd;  // fl(1 / sqrt(d))
 };
 
 // ------------------------------------------------------------- PTX helpers
@@ -401,7 +400,7 @@ __global__ void __launch_bounds__(THREADS, 1)
             screen_init(sr);
             int32_t best = 0x7fffffff, besti = 0x7fffffff;
             float fbest = INFINITY;
-            float a2 = 0.0f, rnx2 = 0.0f, rF = 0.0f, rpc = 0.0f;
+            float a2 = 0.0f, rnx2 = 0.0f, rf2 = 0.0f, rpc = 0.0f;
             int32_t nxr = 0;
             if (MODE == MODE_SCREEN) {
                 a2 = valid ? 2.0f * p.xinfo[row].x : 0.0f;
@@ -409,7 +408,7 @@ __global__ void __launch_bounds__(THREADS, 1)
                 nxr = valid ? p.nx[row] : 0;
             } else {
                 rnx2 = valid ? p.nx2[row] : 0.0f;
-                rF = valid ? p.F[row] : 0.0f;
+                rf2 = valid ? __fmul_rn(-2.0f, p.F[row]) : 0.0f;  // exact
                 rpc = valid ? (float)(2 * p.popx[row] - p.d) : 0.0f;
             }
             for (int ct = 0; ct < p.nct; ++ct, ++job) {
@@ -476,7 +475,8 @@ __global__ void __launch_bounds__(THREADS, 1)
                         }
                     } else {
                         // Eq. final:rabitq in Eq. rabitq_l2 in the library's fixed
-                        // fp32 order, scalar IEEE operations only (packed f32x2
+                        // fp32 order (u = fma(sd, 2P - sum ybar, bd pc),
+                        // est = fma(-2F, u, nx2 + ny2)), scalar IEEE operations (packed f32x2
                         // sequences were measured not to reproduce it).  The e4m3
                         // accumulator carries a small non-integer error (~2^-12),
                         // so P is its nearest integer; 2P - sum ybar is exact.
@@ -497,12 +497,8 @@ __global__ void __launch_bounds__(THREADS, 1)
                                 for (int o = 0; o < 2; ++o) {
                                     const float P = rintf(__uint_as_float(v[i + o]));
                                     const float qv = __fmaf_rn(2.0f, P, nq[o]);  // exact
-                                    const float t1 = __fmul_rn(ss[o], qv);
-                                    const float t2 = __fmul_rn(bb[o], rpc);
-                                    const float ip = __fmul_rn(__fadd_rn(t1, t2), p.isd);
-                                    const float nn = __fadd_rn(rnx2, ny[o]);
-                                    const float fi = __fmul_rn(rF, ip);
-                                    const float est = __fsub_rn(nn, __fmul_rn(2.0f, fi));
+                                    const float u = __fmaf_rn(ss[o], qv, __fmul_rn(bb[o], rpc));
+                                    const float est = __fmaf_rn(rf2, u, __fadd_rn(rnx2, ny[o]));
                                     if (est < gb[g]) {
                                         gb[g] = est;
                                         gi[g] = j0 + i + o;
@@ -780,7 +776,7 @@ __global__ void screen_prep_rbq1_kernel(const uint32_t *__restrict__ codes, int6
 }
 
 // Per-centroid estimator terms -> column-pair records for the tensor
-// epilogue: bs[p] = (b x2, s x2), qn[p] = (-sum ybar x2, ||c - m||^2 x2);
+// epilogue: bs[p] = (bd x2, sd x2), qn[p] = (-sum ybar x2, ||c - m||^2 x2);
 // columns past k get ||c - m||^2 = +inf (never the nearest).
 __global__ void pack_rbq1_pairs_kernel(const Rbq1CInfo *__restrict__ info, int k, int kp,
                                        float4 *__restrict__ bs, float4 *__restrict__ qn) {
@@ -792,8 +788,8 @@ __global__ void pack_rbq1_pairs_kernel(const Rbq1CInfo *__restrict__ info, int k
         const int j = 2 * pp + o;
         if (j < k) {
             const Rbq1CInfo in = info[j];
-            b[o] = in.b;
-            sc[o] = in.s;
+            b[o] = in.bd;
+            sc[o] = in.sd;
             q[o] = -(float)in.sumy;
             n2[o] = in.ny2;
         } else {
@@ -1218,7 +1214,6 @@ int tc_assign_rbq1(const skm_data *x, const float *C, int k, int32_t *assign, fl
     p.F = x->F;
     p.popx = x->popx;
     p.d = d;
-    p.isd = (float)(1.0 / sqrt((double)d));
     SKM_TRY(launch_tc<MODE_RBQ1>(v.xs, n, dp, d, b.cs, k, p, st));
     add_stats_kernel<<<1, 1, 0, st>>>(b.counters, b.stats);
     SKM_CUDA_TRY(launched());

@@ -305,13 +305,51 @@ __device__ __forceinline__ float rbq1_finish(int64_t T, int64_t U, int64_t cnt, 
     return __double2float_rn(__dadd_rn((double)m, v));
 }
 
-// Warp w takes members w, w + 8, ...; word t of a member is loaded by lane t
-// and broadcast; lane l owns dimension 32 t + l of every word t.  Per-warp
-// int64 partials are combined with shared-memory atomics (exact).
+// Fixed-point weights Fq = rint(F 2^e), once per update call.
+__global__ void rbq1_fq_kernel(const float *__restrict__ F, int64_t n, int e,
+                               int64_t *__restrict__ fq) {
+    const double pow2 = ldexp(1.0, e);
+    for (int64_t t = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; t < n;
+         t += (int64_t)gridDim.x * blockDim.x)
+        fq[t] = __double2ll_rn(__dmul_rn((double)F[t], pow2));
+}
+
+cudaError_t launch_rbq1_fq(const float *F, int64_t n, int e, int64_t *fq, cudaStream_t st) {
+    int64_t blocks = (n + 255) / 256;
+    if (blocks > 152 * 8) blocks = 152 * 8;
+    if (blocks < 1) blocks = 1;
+    rbq1_fq_kernel<<<(int)blocks, 256, 0, st>>>(F, n, e, fq);
+    return launched();
+}
+
+// Warp w takes members w, w + 8, ...; the member's code words are read as
+// warp-wide broadcasts (128-bit when the row stride allows) and lane l owns
+// dimension 32 t + l of every word t.  Per-warp int64 partials are combined
+// with shared-memory atomics (exact, order-independent).
 constexpr int RB_WORDS = 32;  // words per pass (1024 dimensions)
 
+template <bool VEC4>
+__device__ __forceinline__ void rb_load_words(const uint32_t *__restrict__ row, int nw,
+                                              uint32_t (&w)[RB_WORDS]) {
+    if (VEC4) {
+#pragma unroll
+        for (int q = 0; q < RB_WORDS / 4; ++q) {
+            uint4 v = make_uint4(0u, 0u, 0u, 0u);
+            if (4 * q < nw) v = __ldg(reinterpret_cast<const uint4 *>(row) + q);
+            w[4 * q] = v.x;
+            w[4 * q + 1] = v.y;
+            w[4 * q + 2] = v.z;
+            w[4 * q + 3] = v.w;
+        }
+    } else {
+#pragma unroll
+        for (int t = 0; t < RB_WORDS; ++t) w[t] = (t < nw) ? __ldg(row + t) : 0u;
+    }
+}
+
+template <bool VEC4>
 __global__ void __launch_bounds__(SEG_THREADS) segsum_rbq1_kernel(
-    const uint32_t *__restrict__ codes, const float *__restrict__ F, int d,
+    const uint32_t *__restrict__ codes, const int64_t *__restrict__ fqs, int d,
     const float *__restrict__ m, int e, const int32_t *__restrict__ perm,
     const int64_t *__restrict__ offsets, float *__restrict__ C, int64_t *__restrict__ partial) {
     __shared__ unsigned long long tot[RB_WORDS * 32];
@@ -322,7 +360,6 @@ __global__ void __launch_bounds__(SEG_THREADS) segsum_rbq1_kernel(
     if (cnt == 0) return;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int W = (d + 31) >> 5;
-    const double pow2 = ldexp(1.0, e);
     const double pow2m = ldexp(1.0, -e);
     const double isd = __ddiv_rn(1.0, __dsqrt_rn((double)d));
     for (int w0 = 0; w0 < W; w0 += RB_WORDS) {
@@ -336,14 +373,13 @@ __global__ void __launch_bounds__(SEG_THREADS) segsum_rbq1_kernel(
         int64_t usum = 0;
         for (int64_t q = lo + warp; q < hi; q += SEG_WARPS) {
             const int64_t p = perm[q];
-            const int64_t fq = __double2ll_rn(__dmul_rn((double)__ldg(F + p), pow2));
+            const int64_t fq = __ldg(fqs + p);
             usum += fq;
-            const uint32_t mine = (lane < nw) ? __ldg(codes + p * W + w0 + lane) : 0u;
+            uint32_t wd[RB_WORDS];
+            rb_load_words<VEC4>(codes + p * W + w0, nw, wd);
 #pragma unroll
-            for (int t = 0; t < RB_WORDS; ++t) {
-                const uint32_t word = __shfl_sync(0xffffffffu, mine, t);
-                if ((word >> lane) & 1u) acc[t] += fq;
-            }
+            for (int t = 0; t < RB_WORDS; ++t)
+                if ((wd[t] >> lane) & 1u) acc[t] += fq;
         }
 #pragma unroll
         for (int t = 0; t < RB_WORDS; ++t)
@@ -365,11 +401,16 @@ __global__ void __launch_bounds__(SEG_THREADS) segsum_rbq1_kernel(
     }
 }
 
-cudaError_t launch_segsum_rbq1(const uint32_t *codes, const float *F, int d, const float *m,
+cudaError_t launch_segsum_rbq1(const uint32_t *codes, const int64_t *fq, int d, const float *m,
                                int e, const int32_t *perm, const int64_t *offsets, int k,
                                float *C_inout, int64_t *partial, cudaStream_t st) {
-    segsum_rbq1_kernel<<<k, SEG_THREADS, 0, st>>>(codes, F, d, m, e, perm, offsets, C_inout,
-                                                  partial);
+    const int W = (d + 31) >> 5;
+    if (W % 4 == 0 && ((uintptr_t)codes & 15) == 0)
+        segsum_rbq1_kernel<true><<<k, SEG_THREADS, 0, st>>>(codes, fq, d, m, e, perm, offsets,
+                                                            C_inout, partial);
+    else
+        segsum_rbq1_kernel<false><<<k, SEG_THREADS, 0, st>>>(codes, fq, d, m, e, perm, offsets,
+                                                             C_inout, partial);
     return launched();
 }
 

@@ -115,6 +115,7 @@ static void plan_assign(const skm_data *x, int k, Carver &cv, AssignBufs &b) {
 struct UpdateBufs {
     int32_t *counts32 = nullptr, *cursor = nullptr, *perm = nullptr;
     int64_t *offsets = nullptr;
+    int64_t *fq = nullptr;  // RBQ1: fixed-point weights round(F 2^e)
 };
 
 static void plan_update(const skm_data *x, int k, Carver &cv, UpdateBufs &b) {
@@ -122,6 +123,7 @@ static void plan_update(const skm_data *x, int k, Carver &cv, UpdateBufs &b) {
     b.cursor = cv.take<int32_t>(k);
     b.offsets = cv.take<int64_t>((size_t)k + 1);
     b.perm = cv.take<int32_t>(x->n);
+    if (x->repr == SKM_REPR_RBQ1) b.fq = cv.take<int64_t>(x->n);
 }
 
 struct FitBufs {
@@ -224,7 +226,8 @@ static int do_update(const skm_data *x, const int32_t *assign, int k, void *C, i
                                        st));
         break;
     case SKM_REPR_RBQ1:
-        SKM_CUDA_TRY(launch_segsum_rbq1(static_cast<const uint32_t *>(x->x), x->F, d, x->m, e,
+        SKM_CUDA_TRY(launch_rbq1_fq(x->F, n, e, b.fq, st));
+        SKM_CUDA_TRY(launch_segsum_rbq1(static_cast<const uint32_t *>(x->x), b.fq, d, x->m, e,
                                         b.perm, b.offsets, k, static_cast<float *>(C),
                                         static_cast<int64_t *>(partial), st));
         break;

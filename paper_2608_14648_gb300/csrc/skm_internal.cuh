@@ -3,6 +3,7 @@
 // here; every launcher returns cudaGetLastError() of its launch.
 #pragma once
 
+#include <math.h>
 #include <cuda_runtime.h>
 #include <cuda_bf16.h>
 #include <stdint.h>
@@ -55,10 +56,11 @@ inline int words_of(int d) { return (d + 31) / 32; }
 inline int64_t cdiv(int64_t a, int64_t b) { return (a + b - 1) / b; }
 
 // Per-centroid terms of the RBQ1 estimator (Eq. final:rabitq), one record
-// per centroid: SQ4 bias b, scale s, sum of codes, ||c - m||^2.
+// per centroid: SQ4 bias and scale multiplied by fl(1/sqrt(d)) (bd = b isd,
+// sd = s isd), the sum of codes, ||c - m||^2.
 struct Rbq1CInfo {
-    float b;
-    float s;
+    float bd;
+    float sd;
     int32_t sumy;
     float ny2;
 };
@@ -84,6 +86,8 @@ cudaError_t launch_rbq1_exponent(const float *F, int64_t n, unsigned int *maxbit
 // centroid preparation
 cudaError_t launch_rbq1_cprep(const float *C, int k, int d, const float *m, uint4 *planes,
                               Rbq1CInfo *info, cudaStream_t st);
+// fl(1 / sqrt(d)) as both sides of the estimator use it
+inline float rbq1_isd(int d) { return (float)(1.0 / sqrt((double)d)); }
 cudaError_t launch_rbq1_cprep_tc(const float *C, int k, int d, const float *m, uint8_t *yq, int dq,
                                  Rbq1CInfo *info, cudaStream_t st);
 cudaError_t launch_row_sqnorm_u8(const uint8_t *codes, int64_t n, int d, int32_t *out,
@@ -121,7 +125,8 @@ cudaError_t launch_segsum_float(const void *X, int x_is_bf16, int d, const int32
 cudaError_t launch_segsum_sq8(const uint8_t *X, int d, const int32_t *perm,
                               const int64_t *offsets, int k, uint8_t *C_inout, int64_t *partial,
                               cudaStream_t st);
-cudaError_t launch_segsum_rbq1(const uint32_t *codes, const float *F, int d, const float *m,
+cudaError_t launch_rbq1_fq(const float *F, int64_t n, int e, int64_t *fq, cudaStream_t st);
+cudaError_t launch_segsum_rbq1(const uint32_t *codes, const int64_t *fq, int d, const float *m,
                                int e, const int32_t *perm, const int64_t *offsets, int k,
                                float *C_inout, int64_t *partial, cudaStream_t st);
 cudaError_t launch_finalize_float(const double *partial, const int64_t *counts, int k, int d,

@@ -236,6 +236,17 @@ def test_rbq1_estimator_matches_direct_sum_and_is_exact_on_grid():
     np.testing.assert_allclose(est, true, rtol=2e-6, atol=2e-5)
 
 
+def test_blocked_sum_of_squares_is_the_sum_of_squares():
+    r = _rng(17)
+    for d in (1, 31, 32, 33, 768, 1000):
+        v = r.standard_normal(d).astype(np.float32)
+        exact = math.fsum(float(x) * float(x) for x in v)
+        assert math.isclose(oracle.sumsq_blocked(v), exact, rel_tol=1e-14)
+    # order matters only through rounding: a permutation inside a block changes nothing
+    v = np.arange(32, dtype=np.float32)
+    assert oracle.sumsq_blocked(v) == sum(float(x) ** 2 for x in v)
+
+
 def test_rbq1_hand_worked_d32_example():
     g = json.load(open(os.path.join(GOLDEN, "rbq1_d32_hand_example.json")))
     d = g["d"]
