@@ -2,9 +2,11 @@
 // Section 3.1): a sort-by-cluster segmented reduction.
 //   1. histogram of assignments (shared-memory privatised counters),
 //   2. exclusive scan -> per-cluster offsets,
-//   3. scatter point ids into cluster-contiguous order,
-//   4. one CTA per cluster sums its members' rows (coalesced row reads) and
-//      finalises the centroid (or adds into caller partial sums).
+//   3. scatter point ids (and their cluster) into cluster-contiguous order,
+//   4. fp32/bf16 and 1-bit: warps take equal runs of the sorted order and
+//      flush per-cluster register sums with global atomics (load balanced
+//      whatever the cluster sizes); SQ8: one CTA per cluster;
+//   5. finalise: divide by the counts (or add into caller partial sums).
 // Integer representations accumulate in int64 and are exact, so their result
 // does not depend on the member order produced by the scatter.
 #include "skm_internal.cuh"
@@ -94,30 +96,29 @@ cudaError_t launch_scan_offsets(const int32_t *counts32, int k, int64_t *offsets
 // ------------------------------------------------------------------ scatter
 __global__ void scatter_kernel(const int32_t *__restrict__ assign, int64_t n, int k,
                                const int64_t *__restrict__ offsets, int32_t *__restrict__ cursor,
-                               int32_t *__restrict__ perm) {
+                               int32_t *__restrict__ perm, int32_t *__restrict__ scl) {
     for (int64_t t = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; t < n;
          t += (int64_t)gridDim.x * blockDim.x) {
         const int a = assign[t];
         if (a < 0 || a >= k) continue;  // skipped consistently with the histogram
         const int pos = atomicAdd(&cursor[a], 1);
         perm[offsets[a] + pos] = (int32_t)t;
+        if (scl) scl[offsets[a] + pos] = a;
     }
 }
 
 cudaError_t launch_scatter(const int32_t *assign, int64_t n, int k, const int64_t *offsets,
-                           int32_t *cursor, int32_t *perm, cudaStream_t st) {
+                           int32_t *cursor, int32_t *perm, int32_t *scl, cudaStream_t st) {
     if (n == 0) return cudaSuccess;
     int64_t blocks = (n + 255) / 256;
     if (blocks > 152 * 8) blocks = 152 * 8;
-    scatter_kernel<<<(unsigned)blocks, 256, 0, st>>>(assign, n, k, offsets, cursor, perm);
+    scatter_kernel<<<(unsigned)blocks, 256, 0, st>>>(assign, n, k, offsets, cursor, perm, scl);
     return launched();
 }
 
-// ------------------------------------------------------ segmented sums: float
-// One CTA per cluster, 8 warps; warp w takes members w, w + 8, ... (two rows
-// in flight), lane l accumulates 16-byte column groups l, l + 32, ... of a
-// 1024-element column chunk.  Warp partials meet in shared memory and are
-// summed in warp order.
+// ------------------------------------------------------ row loads for the sums
+// Lane l reads 16-byte column groups l, l + 32, ... of a 1024-element column
+// chunk of a point row (fp32 or bf16), zero past d.
 constexpr int SEG_WARPS = 8;
 constexpr int SEG_THREADS = SEG_WARPS * 32;
 constexpr int SEG_CHUNK = 1024;  // columns per pass (float: 8 float4 per lane)
@@ -159,65 +160,6 @@ __device__ __forceinline__ void seg_load8(const void *X, int64_t p, int d, int c
         v[4 * g + 2] = f.z;
         v[4 * g + 3] = f.w;
     }
-}
-
-template <bool BF16>
-__global__ void __launch_bounds__(SEG_THREADS) segsum_float_kernel(
-    const void *__restrict__ Xv, int d, const int32_t *__restrict__ perm,
-    const int64_t *__restrict__ offsets, float *__restrict__ C, double *__restrict__ partial) {
-    __shared__ float red[SEG_WARPS][SEG_CHUNK];
-    const int j = blockIdx.x;
-    const int64_t lo = offsets[j], hi = offsets[j + 1];
-    const int64_t cnt = hi - lo;
-    if (cnt == 0) return;  // empty cluster keeps its centroid / adds nothing
-    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    for (int c0 = 0; c0 < d; c0 += SEG_CHUNK) {
-        float acc[SEG_CHUNK / 32];
-#pragma unroll
-        for (int t = 0; t < SEG_CHUNK / 32; ++t) acc[t] = 0.0f;
-        int64_t q = lo + warp;
-        for (; q + SEG_WARPS < hi; q += 2 * SEG_WARPS) {
-            float v0[SEG_CHUNK / 32], v1[SEG_CHUNK / 32];
-            seg_load8<BF16>(Xv, perm[q], d, c0, lane, v0);
-            seg_load8<BF16>(Xv, perm[q + SEG_WARPS], d, c0, lane, v1);
-#pragma unroll
-            for (int t = 0; t < SEG_CHUNK / 32; ++t) acc[t] += v0[t] + v1[t];
-        }
-        if (q < hi) {
-            float v0[SEG_CHUNK / 32];
-            seg_load8<BF16>(Xv, perm[q], d, c0, lane, v0);
-#pragma unroll
-            for (int t = 0; t < SEG_CHUNK / 32; ++t) acc[t] += v0[t];
-        }
-        __syncthreads();
-#pragma unroll
-        for (int g = 0; g < SEG_CHUNK / 128; ++g)
-#pragma unroll
-            for (int u = 0; u < 4; ++u) red[warp][4 * (lane + 32 * g) + u] = acc[4 * g + u];
-        __syncthreads();
-        for (int t = threadIdx.x; t < SEG_CHUNK; t += SEG_THREADS) {
-            const int i = c0 + t;
-            if (i >= d) break;
-            float s = 0.0f;
-#pragma unroll
-            for (int w = 0; w < SEG_WARPS; ++w) s += red[w][t];
-            if (partial)
-                partial[(int64_t)j * d + i] += (double)s;
-            else
-                C[(int64_t)j * d + i] = __fdiv_rn(s, (float)cnt);
-        }
-    }
-}
-
-cudaError_t launch_segsum_float(const void *X, int x_is_bf16, int d, const int32_t *perm,
-                                const int64_t *offsets, int k, float *C_inout, double *partial,
-                                cudaStream_t st) {
-    if (x_is_bf16)
-        segsum_float_kernel<true><<<k, SEG_THREADS, 0, st>>>(X, d, perm, offsets, C_inout, partial);
-    else
-        segsum_float_kernel<false><<<k, SEG_THREADS, 0, st>>>(X, d, perm, offsets, C_inout,
-                                                              partial);
-    return launched();
 }
 
 // ------------------------------------------------------- segmented sums: SQ8
@@ -322,95 +264,175 @@ cudaError_t launch_rbq1_fq(const float *F, int64_t n, int e, int64_t *fq, cudaSt
     return launched();
 }
 
-// Warp w takes members w, w + 8, ...; the member's code words are read as
-// warp-wide broadcasts (128-bit when the row stride allows) and lane l owns
-// dimension 32 t + l of every word t.  Per-warp int64 partials are combined
-// with shared-memory atomics (exact, order-independent).
-constexpr int RB_WORDS = 32;  // words per pass (1024 dimensions)
+constexpr int RB_WORDS = 32;  // code words per pass (1024 dimensions)
 
-template <bool VEC4>
-__device__ __forceinline__ void rb_load_words(const uint32_t *__restrict__ row, int nw,
-                                              uint32_t (&w)[RB_WORDS]) {
-    if (VEC4) {
+// -------------------------------------------- chunked segmented sums (load balanced)
+// Warps take CH_ROWS consecutive members of the cluster-sorted order, so
+// every warp has the same work whatever the cluster sizes.  A warp adds its
+// rows into register accumulators and flushes them with global atomics into
+// the cluster's accumulator whenever the cluster changes (and at the end).
+// The member count of the sorted order is offsets[k].
+constexpr int CH_WARPS = 8;
+constexpr int CH_ROWS = 128;
+
+// fp32 / bf16 points -> float or double accumulators S[k][d].
+template <bool BF16, typename ACC>
+__global__ void __launch_bounds__(CH_WARPS * 32) chunk_sum_float_kernel(
+    const void *__restrict__ Xv, int d, const int32_t *__restrict__ perm,
+    const int32_t *__restrict__ scl, const int64_t *__restrict__ offsets, int k,
+    ACC *__restrict__ S, int64_t stride) {
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int64_t nval = offsets[k];
+    const int64_t q0 = ((int64_t)blockIdx.x * CH_WARPS + warp) * CH_ROWS;
+    if (q0 >= nval) return;
+    const int64_t q1 = min(nval, q0 + CH_ROWS);
+    for (int c0 = 0; c0 < d; c0 += SEG_CHUNK) {
+        float acc[SEG_CHUNK / 32];
 #pragma unroll
-        for (int q = 0; q < RB_WORDS / 4; ++q) {
-            uint4 v = make_uint4(0u, 0u, 0u, 0u);
-            if (4 * q < nw) v = __ldg(reinterpret_cast<const uint4 *>(row) + q);
-            w[4 * q] = v.x;
-            w[4 * q + 1] = v.y;
-            w[4 * q + 2] = v.z;
-            w[4 * q + 3] = v.w;
+        for (int t = 0; t < SEG_CHUNK / 32; ++t) acc[t] = 0.0f;
+        int cur = scl[q0];
+        auto flush = [&](int c) {
+#pragma unroll
+            for (int g = 0; g < SEG_CHUNK / 128; ++g)
+#pragma unroll
+                for (int u = 0; u < 4; ++u) {
+                    const int col = c0 + 4 * (lane + 32 * g) + u;
+                    if (col < d) atomicAdd(S + (int64_t)c * stride + col, (ACC)acc[4 * g + u]);
+                    acc[4 * g + u] = 0.0f;
+                }
+        };
+        int64_t q = q0;
+        for (; q + 1 < q1; q += 2) {
+            const int ca = scl[q], cb = scl[q + 1];
+            float v0[SEG_CHUNK / 32], v1[SEG_CHUNK / 32];
+            seg_load8<BF16>(Xv, perm[q], d, c0, lane, v0);
+            seg_load8<BF16>(Xv, perm[q + 1], d, c0, lane, v1);
+            if (ca != cur) {
+                flush(cur);
+                cur = ca;
+            }
+#pragma unroll
+            for (int t = 0; t < SEG_CHUNK / 32; ++t) acc[t] += v0[t];
+            if (cb != cur) {
+                flush(cur);
+                cur = cb;
+            }
+#pragma unroll
+            for (int t = 0; t < SEG_CHUNK / 32; ++t) acc[t] += v1[t];
         }
-    } else {
+        if (q < q1) {
+            const int ca = scl[q];
+            float v0[SEG_CHUNK / 32];
+            seg_load8<BF16>(Xv, perm[q], d, c0, lane, v0);
+            if (ca != cur) {
+                flush(cur);
+                cur = ca;
+            }
 #pragma unroll
-        for (int t = 0; t < RB_WORDS; ++t) w[t] = (t < nw) ? __ldg(row + t) : 0u;
+            for (int t = 0; t < SEG_CHUNK / 32; ++t) acc[t] += v0[t];
+        }
+        flush(cur);
     }
 }
 
-template <bool VEC4>
-__global__ void __launch_bounds__(SEG_THREADS) segsum_rbq1_kernel(
+// 1-bit codes -> int64 accumulators T[k][d+1] (column d holds U = sum Fq).
+__global__ void __launch_bounds__(CH_WARPS * 32) chunk_sum_rbq1_kernel(
     const uint32_t *__restrict__ codes, const int64_t *__restrict__ fqs, int d,
-    const float *__restrict__ m, int e, const int32_t *__restrict__ perm,
-    const int64_t *__restrict__ offsets, float *__restrict__ C, int64_t *__restrict__ partial) {
-    __shared__ unsigned long long tot[RB_WORDS * 32];
-    __shared__ unsigned long long utot;
-    const int j = blockIdx.x;
-    const int64_t lo = offsets[j], hi = offsets[j + 1];
-    const int64_t cnt = hi - lo;
-    if (cnt == 0) return;
+    const int32_t *__restrict__ perm, const int32_t *__restrict__ scl,
+    const int64_t *__restrict__ offsets, int k, unsigned long long *__restrict__ T) {
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int64_t nval = offsets[k];
+    const int64_t q0 = ((int64_t)blockIdx.x * CH_WARPS + warp) * CH_ROWS;
+    if (q0 >= nval) return;
+    const int64_t q1 = min(nval, q0 + CH_ROWS);
     const int W = (d + 31) >> 5;
-    const double pow2m = ldexp(1.0, -e);
-    const double isd = __ddiv_rn(1.0, __dsqrt_rn((double)d));
     for (int w0 = 0; w0 < W; w0 += RB_WORDS) {
         const int nw = min(RB_WORDS, W - w0);
-        for (int t = threadIdx.x; t < RB_WORDS * 32; t += SEG_THREADS) tot[t] = 0ull;
-        if (threadIdx.x == 0 && w0 == 0) utot = 0ull;  // U is summed in the first pass only
-        __syncthreads();
         int64_t acc[RB_WORDS];
 #pragma unroll
         for (int t = 0; t < RB_WORDS; ++t) acc[t] = 0;
         int64_t usum = 0;
-        for (int64_t q = lo + warp; q < hi; q += SEG_WARPS) {
+        int cur = scl[q0];
+        auto flush = [&](int c) {
+#pragma unroll
+            for (int t = 0; t < RB_WORDS; ++t) {
+                const int col = 32 * (w0 + t) + lane;
+                if (t < nw && col < d && acc[t])
+                    atomicAdd(T + (int64_t)c * (d + 1) + col, (unsigned long long)acc[t]);
+                acc[t] = 0;
+            }
+            if (w0 == 0 && lane == 0 && usum) atomicAdd(T + (int64_t)c * (d + 1) + d, (unsigned long long)usum);
+            usum = 0;
+        };
+        for (int64_t q = q0; q < q1; ++q) {
+            const int c = scl[q];
             const int64_t p = perm[q];
             const int64_t fq = __ldg(fqs + p);
+            const uint32_t mine = (lane < nw) ? __ldg(codes + p * W + w0 + lane) : 0u;
+            if (c != cur) {
+                flush(cur);
+                cur = c;
+            }
             usum += fq;
-            uint32_t wd[RB_WORDS];
-            rb_load_words<VEC4>(codes + p * W + w0, nw, wd);
 #pragma unroll
-            for (int t = 0; t < RB_WORDS; ++t)
-                if ((wd[t] >> lane) & 1u) acc[t] += fq;
+            for (int t = 0; t < RB_WORDS; ++t) {
+                const uint32_t word = __shfl_sync(0xffffffffu, mine, t);
+                if ((word >> lane) & 1u) acc[t] += fq;
+            }
         }
-#pragma unroll
-        for (int t = 0; t < RB_WORDS; ++t)
-            if (t < nw && acc[t]) atomicAdd(&tot[32 * t + lane], (unsigned long long)acc[t]);
-        if (lane == 0 && w0 == 0) atomicAdd(&utot, (unsigned long long)usum);
-        __syncthreads();
-        const int64_t U = (int64_t)utot;
-        for (int t = threadIdx.x; t < nw * 32; t += SEG_THREADS) {
-            const int i = 32 * w0 + t;
-            if (i >= d) continue;
-            const int64_t T = (int64_t)tot[t];
-            if (partial)
-                partial[(int64_t)j * (d + 1) + i] += T;
-            else
-                C[(int64_t)j * d + i] = rbq1_finish(T, U, cnt, m[i], pow2m, isd);
-        }
-        if (partial && w0 == 0 && threadIdx.x == 0) partial[(int64_t)j * (d + 1) + d] += U;
-        __syncthreads();
+        flush(cur);
     }
 }
 
-cudaError_t launch_segsum_rbq1(const uint32_t *codes, const int64_t *fq, int d, const float *m,
-                               int e, const int32_t *perm, const int64_t *offsets, int k,
-                               float *C_inout, int64_t *partial, cudaStream_t st) {
-    const int W = (d + 31) >> 5;
-    if (W % 4 == 0 && ((uintptr_t)codes & 15) == 0)
-        segsum_rbq1_kernel<true><<<k, SEG_THREADS, 0, st>>>(codes, fq, d, m, e, perm, offsets,
-                                                            C_inout, partial);
-    else
-        segsum_rbq1_kernel<false><<<k, SEG_THREADS, 0, st>>>(codes, fq, d, m, e, perm, offsets,
-                                                             C_inout, partial);
+static unsigned chunk_blocks(int64_t n) {
+    const int64_t per = (int64_t)CH_WARPS * CH_ROWS;
+    int64_t b = (n + per - 1) / per;
+    return (unsigned)(b < 1 ? 1 : b);
+}
+
+cudaError_t launch_chunk_sum_float(const void *X, int x_is_bf16, int64_t n, int d,
+                                   const int32_t *perm, const int32_t *scl,
+                                   const int64_t *offsets, int k, float *S_f, double *S_d,
+                                   cudaStream_t st) {
+    if (n == 0) return cudaSuccess;
+    const unsigned g = chunk_blocks(n);
+    if (S_d) {
+        if (x_is_bf16)
+            chunk_sum_float_kernel<true, double><<<g, CH_WARPS * 32, 0, st>>>(X, d, perm, scl, offsets, k, S_d, d);
+        else
+            chunk_sum_float_kernel<false, double><<<g, CH_WARPS * 32, 0, st>>>(X, d, perm, scl, offsets, k, S_d, d);
+    } else {
+        if (x_is_bf16)
+            chunk_sum_float_kernel<true, float><<<g, CH_WARPS * 32, 0, st>>>(X, d, perm, scl, offsets, k, S_f, d);
+        else
+            chunk_sum_float_kernel<false, float><<<g, CH_WARPS * 32, 0, st>>>(X, d, perm, scl, offsets, k, S_f, d);
+    }
+    return launched();
+}
+
+cudaError_t launch_chunk_sum_rbq1(const uint32_t *codes, const int64_t *fq, int64_t n, int d,
+                                  const int32_t *perm, const int32_t *scl, const int64_t *offsets,
+                                  int k, int64_t *T, cudaStream_t st) {
+    if (n == 0) return cudaSuccess;
+    chunk_sum_rbq1_kernel<<<chunk_blocks(n), CH_WARPS * 32, 0, st>>>(
+        codes, fq, d, perm, scl, offsets, k, reinterpret_cast<unsigned long long *>(T));
+    return launched();
+}
+
+// fp32 sums -> centroids (clusters without members keep theirs)
+__global__ void finalize_float32_kernel(const float *__restrict__ S,
+                                        const int64_t *__restrict__ counts, int k, int d,
+                                        float *__restrict__ C) {
+    const int64_t t = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
+    if (t >= (int64_t)k * d) return;
+    const int64_t c = counts[t / d];
+    if (c > 0) C[t] = __fdiv_rn(S[t], (float)c);
+}
+
+cudaError_t launch_finalize_float32(const float *S, const int64_t *counts, int k, int d,
+                                    float *C_inout, cudaStream_t st) {
+    const int64_t tot = (int64_t)k * d;
+    finalize_float32_kernel<<<(unsigned)((tot + 255) / 256), 256, 0, st>>>(S, counts, k, d, C_inout);
     return launched();
 }
 

@@ -113,9 +113,11 @@ static void plan_assign(const skm_data *x, int k, Carver &cv, AssignBufs &b) {
 }
 
 struct UpdateBufs {
-    int32_t *counts32 = nullptr, *cursor = nullptr, *perm = nullptr;
+    int32_t *counts32 = nullptr, *cursor = nullptr, *perm = nullptr, *scl = nullptr;
     int64_t *offsets = nullptr;
-    int64_t *fq = nullptr;  // RBQ1: fixed-point weights round(F 2^e)
+    int64_t *fq = nullptr;    // RBQ1: fixed-point weights round(F 2^e)
+    float *sumf = nullptr;    // F32/BF16: cluster sums [k][d]
+    int64_t *sumi = nullptr;  // RBQ1: cluster sums [k][d + 1]
 };
 
 static void plan_update(const skm_data *x, int k, Carver &cv, UpdateBufs &b) {
@@ -123,7 +125,12 @@ static void plan_update(const skm_data *x, int k, Carver &cv, UpdateBufs &b) {
     b.cursor = cv.take<int32_t>(k);
     b.offsets = cv.take<int64_t>((size_t)k + 1);
     b.perm = cv.take<int32_t>(x->n);
-    if (x->repr == SKM_REPR_RBQ1) b.fq = cv.take<int64_t>(x->n);
+    b.scl = cv.take<int32_t>(x->n);
+    if (x->repr == SKM_REPR_RBQ1) {
+        b.fq = cv.take<int64_t>(x->n);
+        b.sumi = cv.take<int64_t>((size_t)k * (x->d + 1));
+    }
+    if (x->repr == SKM_REPR_F32 || x->repr == SKM_REPR_BF16) b.sumf = cv.take<float>((size_t)k * x->d);
 }
 
 struct FitBufs {
@@ -212,25 +219,36 @@ static int do_update(const skm_data *x, const int32_t *assign, int k, void *C, i
     SKM_CUDA_TRY(launch_histogram(assign, n, k, b.counts32, st));
     SKM_CUDA_TRY(launch_scan_offsets(b.counts32, k, b.offsets, counts, partial ? 1 : 0, st));
     SKM_CUDA_TRY(cudaMemsetAsync(b.cursor, 0, sizeof(int32_t) * (size_t)k, st));
-    SKM_CUDA_TRY(launch_scatter(assign, n, k, b.offsets, b.cursor, b.perm, st));
+    SKM_CUDA_TRY(launch_scatter(assign, n, k, b.offsets, b.cursor, b.perm, b.scl, st));
     switch (x->repr) {
     case SKM_REPR_F32:
     case SKM_REPR_BF16:
-        SKM_CUDA_TRY(launch_segsum_float(x->x, x->repr == SKM_REPR_BF16, d, b.perm, b.offsets, k,
-                                         static_cast<float *>(C), static_cast<double *>(partial),
-                                         st));
+        if (partial) {
+            SKM_CUDA_TRY(launch_chunk_sum_float(x->x, x->repr == SKM_REPR_BF16, n, d, b.perm, b.scl,
+                                                b.offsets, k, nullptr,
+                                                static_cast<double *>(partial), st));
+        } else {
+            SKM_CUDA_TRY(cudaMemsetAsync(b.sumf, 0, sizeof(float) * (size_t)k * d, st));
+            SKM_CUDA_TRY(launch_chunk_sum_float(x->x, x->repr == SKM_REPR_BF16, n, d, b.perm, b.scl,
+                                                b.offsets, k, b.sumf, nullptr, st));
+            SKM_CUDA_TRY(launch_finalize_float32(b.sumf, counts, k, d, static_cast<float *>(C), st));
+        }
         break;
     case SKM_REPR_SQ8:
         SKM_CUDA_TRY(launch_segsum_sq8(static_cast<const uint8_t *>(x->x), d, b.perm, b.offsets, k,
                                        static_cast<uint8_t *>(C), static_cast<int64_t *>(partial),
                                        st));
         break;
-    case SKM_REPR_RBQ1:
+    case SKM_REPR_RBQ1: {
         SKM_CUDA_TRY(launch_rbq1_fq(x->F, n, e, b.fq, st));
-        SKM_CUDA_TRY(launch_segsum_rbq1(static_cast<const uint32_t *>(x->x), b.fq, d, x->m, e,
-                                        b.perm, b.offsets, k, static_cast<float *>(C),
-                                        static_cast<int64_t *>(partial), st));
+        int64_t *T = partial ? static_cast<int64_t *>(partial) : b.sumi;
+        if (!partial) SKM_CUDA_TRY(cudaMemsetAsync(T, 0, sizeof(int64_t) * (size_t)k * (d + 1), st));
+        SKM_CUDA_TRY(launch_chunk_sum_rbq1(static_cast<const uint32_t *>(x->x), b.fq, n, d, b.perm,
+                                           b.scl, b.offsets, k, T, st));
+        if (!partial)
+            SKM_CUDA_TRY(launch_finalize_rbq1(T, counts, k, d, x->m, e, static_cast<float *>(C), st));
         break;
+    }
     }
     return SKM_OK;
 }

@@ -117,18 +117,21 @@ cudaError_t launch_histogram(const int32_t *assign, int64_t n, int k, int32_t *c
 cudaError_t launch_scan_offsets(const int32_t *counts32, int k, int64_t *offsets,
                                 int64_t *counts64_out, int accumulate_counts, cudaStream_t st);
 cudaError_t launch_scatter(const int32_t *assign, int64_t n, int k, const int64_t *offsets,
-                           int32_t *cursor, int32_t *perm, cudaStream_t st);
-// repr: 0 f32, 3 bf16 (float centroids); mode: 0 finalise, 1 accumulate partial
-cudaError_t launch_segsum_float(const void *X, int x_is_bf16, int d, const int32_t *perm,
-                                const int64_t *offsets, int k, float *C_inout, double *partial,
-                                cudaStream_t st);
+                           int32_t *cursor, int32_t *perm, int32_t *scl, cudaStream_t st);
+// load-balanced segmented sums over the cluster-sorted order (global atomics)
+cudaError_t launch_chunk_sum_float(const void *X, int x_is_bf16, int64_t n, int d,
+                                   const int32_t *perm, const int32_t *scl,
+                                   const int64_t *offsets, int k, float *S_f, double *S_d,
+                                   cudaStream_t st);
+cudaError_t launch_chunk_sum_rbq1(const uint32_t *codes, const int64_t *fq, int64_t n, int d,
+                                  const int32_t *perm, const int32_t *scl, const int64_t *offsets,
+                                  int k, int64_t *T, cudaStream_t st);
+cudaError_t launch_finalize_float32(const float *S, const int64_t *counts, int k, int d,
+                                    float *C_inout, cudaStream_t st);
 cudaError_t launch_segsum_sq8(const uint8_t *X, int d, const int32_t *perm,
                               const int64_t *offsets, int k, uint8_t *C_inout, int64_t *partial,
                               cudaStream_t st);
 cudaError_t launch_rbq1_fq(const float *F, int64_t n, int e, int64_t *fq, cudaStream_t st);
-cudaError_t launch_segsum_rbq1(const uint32_t *codes, const int64_t *fq, int d, const float *m,
-                               int e, const int32_t *perm, const int64_t *offsets, int k,
-                               float *C_inout, int64_t *partial, cudaStream_t st);
 cudaError_t launch_finalize_float(const double *partial, const int64_t *counts, int k, int d,
                                   float *C_inout, cudaStream_t st);
 cudaError_t launch_finalize_sq8(const int64_t *partial, const int64_t *counts, int k, int d,
