@@ -476,8 +476,7 @@ __global__ void __launch_bounds__(THREADS, 1)
                     } else {
                         // Eq. final:rabitq in Eq. rabitq_l2 in the library's fixed
                         // fp32 order (u = fma(sd, 2P - sum ybar, bd pc),
-                        // est = fma(-2F, u, nx2 + ny2)), scalar IEEE operations (packed f32x2
-                        // sequences were measured not to reproduce it).  The e4m3
+                        // est = fma(-2F, u, nx2 + ny2)).  The e4m3
                         // accumulator carries a small non-integer error (~2^-12),
                         // so P is its nearest integer; 2P - sum ybar is exact.
                         float gb[4];
@@ -491,18 +490,22 @@ __global__ void __launch_bounds__(THREADS, 1)
                             for (int i = 8 * g; i < 8 * g + 8; i += 2) {
                                 const float4 bs = __ldg(p.rinfo + ((j0 + i) >> 1));
                                 const float4 qn = __ldg(p.rinfoq + ((j0 + i) >> 1));
-                                const float bb[2] = {bs.x, bs.y}, ss[2] = {bs.z, bs.w};
-                                const float nq[2] = {qn.x, qn.y}, ny[2] = {qn.z, qn.w};
-#pragma unroll
-                                for (int o = 0; o < 2; ++o) {
-                                    const float P = rintf(__uint_as_float(v[i + o]));
-                                    const float qv = __fmaf_rn(2.0f, P, nq[o]);  // exact
-                                    const float u = __fmaf_rn(ss[o], qv, __fmul_rn(bb[o], rpc));
-                                    const float est = __fmaf_rn(rf2, u, __fadd_rn(rnx2, ny[o]));
-                                    if (est < gb[g]) {
-                                        gb[g] = est;
-                                        gi[g] = j0 + i + o;
-                                    }
+                                // packed pairs; every product here feeds an explicit fma
+                                // (no separate multiply-add the compiler could fuse)
+                                const float2 P2 = make_float2(rintf(__uint_as_float(v[i])),
+                                                              rintf(__uint_as_float(v[i + 1])));
+                                const float2 qv = ffma2(make_float2(2.0f, 2.0f), P2, make_float2(qn.x, qn.y));
+                                const float2 t = fmul2(make_float2(bs.x, bs.y), make_float2(rpc, rpc));
+                                const float2 u = ffma2(make_float2(bs.z, bs.w), qv, t);
+                                const float2 nn = fadd2(make_float2(rnx2, rnx2), make_float2(qn.z, qn.w));
+                                const float2 est = ffma2(make_float2(rf2, rf2), u, nn);
+                                if (est.x < gb[g]) {
+                                    gb[g] = est.x;
+                                    gi[g] = j0 + i;
+                                }
+                                if (est.y < gb[g]) {
+                                    gb[g] = est.y;
+                                    gi[g] = j0 + i + 1;
                                 }
                             }
                         }
