@@ -1,0 +1,450 @@
+// Streamed segmented sums for the centroid update (Section 2.3 STEP 3; for
+// 1-bit codes the fused decode-average of Section 3.1 "RabitQ").
+//
+// The cluster-sorted member order is cut into runs of RS_ROWS positions and
+// each of the RS_CW consumer warps of a CTA owns one run.  A producer warp
+// gathers the member rows of the CTA's runs with cp.async.bulk (global ->
+// shared, completion counted in bytes on one mbarrier per slot) into a ring
+// of slots per consumer warp, so that tens of rows per SM are in flight
+// without holding them in registers.  A consumer warp adds each row of its run
+// into register accumulators and flushes them into the cluster's global
+// accumulator with atomics whenever the cluster id changes and at the end of
+// the run; every warp has the same number of rows whatever the cluster sizes.
+//
+// Every barrier wait is bounded (2 s of %globaltimer).  A wait that gives up
+// raises *flag (which skm_fit reports as SKM_ERR_TIMEOUT), the warp stops,
+// and the producer waits (bounded again) for the copies it issued before the
+// CTA returns, so no copy lands in the shared memory of a finished CTA.
+#include <algorithm>
+
+#include "skm_internal.cuh"
+
+namespace skm {
+namespace {
+
+constexpr int RS_CW = 8;                      // consumer warps per CTA
+constexpr int RS_THREADS = 32 * (RS_CW + 1);  // + one producer warp
+constexpr int RS_ROWS = 128;                  // sorted positions per consumer warp
+constexpr int RS_MAX_SLOTS = 16;              // ring slots per consumer warp
+constexpr int RS_RING_BYTES = 96 * 1024;      // all rings of a CTA
+constexpr unsigned long long RS_WAIT_NS = 2000000000ull;
+
+__device__ __forceinline__ uint32_t su32(const void *p) { return (uint32_t)__cvta_generic_to_shared(p); }
+__device__ __forceinline__ unsigned long long gtimer() {
+    unsigned long long t;
+    asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+    return t;
+}
+__device__ __forceinline__ void bar_init(uint32_t b, uint32_t count) {
+    asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(b), "r"(count) : "memory");
+}
+__device__ __forceinline__ void bar_arrive(uint32_t b) {
+    asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(b) : "memory");
+}
+__device__ __forceinline__ void bar_arrive_tx(uint32_t b, uint32_t bytes) {
+    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(b), "r"(bytes)
+                 : "memory");
+}
+__device__ __forceinline__ bool bar_try(uint32_t b, uint32_t parity) {
+    uint32_t ok;
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+        "selp.u32 %0, 1, 0, p;\n\t}\n"
+        : "=r"(ok)
+        : "r"(b), "r"(parity)
+        : "memory");
+    return ok != 0;
+}
+// false once the flag is up or the limit has elapsed (the flag is then raised)
+__device__ __forceinline__ bool bar_wait(uint32_t b, uint32_t parity, volatile int32_t *flag) {
+    if (bar_try(b, parity)) return true;
+    const unsigned long long t0 = gtimer();
+    for (uint32_t i = 1;; ++i) {
+        if (bar_try(b, parity)) return true;
+        if ((i & 63) == 0) {
+            if (*flag) return false;
+            if (gtimer() - t0 > RS_WAIT_NS) {
+                *flag = 1;
+                return false;
+            }
+        }
+    }
+}
+// wait with a limit only (used to drain copies already issued)
+__device__ __forceinline__ bool bar_wait_drain(uint32_t b, uint32_t parity) {
+    const unsigned long long t0 = gtimer();
+    while (!bar_try(b, parity))
+        if (gtimer() - t0 > RS_WAIT_NS) return false;
+    return true;
+}
+__device__ __forceinline__ void bulk_g2s(uint32_t dst, const void *src, uint32_t bytes, uint32_t b) {
+    asm volatile(
+        "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(dst),
+        "l"(src), "r"(bytes), "r"(b)
+        : "memory");
+}
+
+__device__ __forceinline__ int run_len(int64_t nval, int64_t q0) {
+    const int64_t r = nval - q0;
+    return r <= 0 ? 0 : (r >= RS_ROWS ? RS_ROWS : (int)r);
+}
+
+// Shared-memory layout of one CTA (ns slots of sb bytes per consumer warp).
+struct RingLayout {
+    int ns, sb;
+    __host__ __device__ size_t ring_bytes() const { return (size_t)RS_CW * ns * sb; }
+    __host__ __device__ size_t bytes() const {
+        return ring_bytes() + (size_t)2 * RS_CW * ns * 8 + (size_t)RS_CW * RS_ROWS * 4 + 2 * RS_CW * 4;
+    }
+};
+
+// Producer and teardown shared by every row type.  A consumer warp calls
+// cons.start(q0, cnt, lane) before the first row of its run (positions q0 ..
+// q0 + cnt - 1), cons.row(i, slot, lane) for its i-th row (in shared memory),
+// and cons.finish(lane) after the last.
+template <typename Consumer>
+__device__ __forceinline__ void ring_run(const uint8_t *__restrict__ rows, uint32_t rb,
+                                         const int32_t *__restrict__ perm, int64_t nval,
+                                         RingLayout L, volatile int32_t *flag, Consumer &cons) {
+    extern __shared__ __align__(128) uint8_t rs_smem[];
+    uint8_t *ring = rs_smem;
+    uint64_t *full = reinterpret_cast<uint64_t *>(rs_smem + L.ring_bytes());
+    uint64_t *empty = full + RS_CW * L.ns;
+    int32_t *sperm = reinterpret_cast<int32_t *>(empty + RS_CW * L.ns);
+    int32_t *issued = sperm + RS_CW * RS_ROWS;
+    int32_t *consumed = issued + RS_CW;
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int64_t qbase = (int64_t)blockIdx.x * RS_CW * RS_ROWS;
+
+    if (threadIdx.x == 0) {
+        for (int i = 0; i < RS_CW * L.ns; ++i) {
+            bar_init(su32(full + i), 1);
+            bar_init(su32(empty + i), 1);
+        }
+        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    }
+    if (threadIdx.x < RS_CW) {
+        issued[threadIdx.x] = 0;
+        consumed[threadIdx.x] = 0;
+    }
+    __syncthreads();
+
+    if (warp == RS_CW) {  // ------------------------------------------ producer
+        for (int i = lane; i < RS_CW * RS_ROWS; i += 32) {
+            const int64_t q = qbase + i;
+            sperm[i] = q < nval ? perm[q] : 0;
+        }
+        __syncwarp();
+        if (lane < RS_CW) {
+            const int w = lane;
+            const int64_t q0 = qbase + (int64_t)w * RS_ROWS;
+            const int cnt = run_len(nval, q0);
+            int i = 0;
+            for (; i < cnt; ++i) {
+                const int s = i % L.ns;
+                const uint32_t ph = (uint32_t)(i / L.ns) & 1u;
+                const uint32_t fb = su32(full + w * L.ns + s);
+                if (!bar_wait(su32(empty + w * L.ns + s), ph ^ 1u, flag)) break;
+                bar_arrive_tx(fb, rb);
+                bulk_g2s(su32(ring + ((size_t)w * L.ns + s) * L.sb),
+                         rows + (size_t)sperm[w * RS_ROWS + i] * rb, rb, fb);
+            }
+            issued[w] = i;
+        }
+    } else {  // ------------------------------------------------------ consumers
+        const int w = warp;
+        const int64_t q0 = qbase + (int64_t)w * RS_ROWS;
+        const int cnt = run_len(nval, q0);
+        int i = 0;
+        if (cnt > 0) {
+            cons.start(q0, cnt, lane);
+            for (; i < cnt; ++i) {
+                const int s = i % L.ns;
+                const uint32_t ph = (uint32_t)(i / L.ns) & 1u;
+                const bool ok = bar_wait(su32(full + w * L.ns + s), ph, flag);
+                if (!__all_sync(0xffffffffu, ok)) break;
+                cons.row(i, ring + ((size_t)w * L.ns + s) * L.sb, lane);
+                __syncwarp();
+                if (lane == 0) bar_arrive(su32(empty + w * L.ns + s));
+            }
+            cons.finish(lane);
+        }
+        if (lane == 0) consumed[w] = i;
+    }
+    __syncthreads();
+    // copies issued but never consumed (only after a wait gave up): let them land
+    if (warp == RS_CW && lane < RS_CW) {
+        const int w = lane;
+        for (int i = consumed[w]; i < issued[w]; ++i) {
+            const int s = i % L.ns;
+            if (!bar_wait_drain(su32(full + w * L.ns + s), (uint32_t)(i / L.ns) & 1u)) break;
+        }
+    }
+}
+
+// ---------------------------------------------------------- fp32 / bf16 rows
+// Lane l holds columns 4 (l + 32 t) .. +3, t < NF.
+template <bool BF16, typename ACC, int NF>
+struct FloatCons {
+    const int32_t *scl;
+    ACC *S;
+    int64_t stride;
+    int d;
+    float acc[4 * NF];
+    int cur;
+    int64_t q0;
+    int clw, cln;  // cluster ids of this and the next 32 positions (lane-held)
+    int cnt;
+    __device__ __forceinline__ void flush(int c, int lane) {
+#pragma unroll
+        for (int t = 0; t < NF; ++t)
+#pragma unroll
+            for (int u = 0; u < 4; ++u) {
+                const int col = 4 * (lane + 32 * t) + u;
+                if (col < d) atomicAdd(S + (int64_t)c * stride + col, (ACC)acc[4 * t + u]);
+                acc[4 * t + u] = 0.0f;
+            }
+    }
+    __device__ __forceinline__ void start(int64_t q0_, int cnt_, int lane) {
+        q0 = q0_;
+        cnt = cnt_;
+#pragma unroll
+        for (int t = 0; t < 4 * NF; ++t) acc[t] = 0.0f;
+        clw = lane < cnt ? __ldg(scl + q0 + lane) : -1;
+        cln = 32 + lane < cnt ? __ldg(scl + q0 + 32 + lane) : -1;
+        cur = __shfl_sync(0xffffffffu, clw, 0);
+    }
+    __device__ __forceinline__ void row(int i, const uint8_t *slot, int lane) {
+        if ((i & 31) == 0 && i > 0) {
+            clw = cln;
+            const int nx = i + 32 + lane;
+            cln = nx < cnt ? __ldg(scl + q0 + nx) : -1;
+        }
+        const int c = __shfl_sync(0xffffffffu, clw, i & 31);
+        if (c != cur) {
+            flush(cur, lane);
+            cur = c;
+        }
+        const int nq = d >> 2;  // float4 groups (d % 4 == 0 on this path)
+#pragma unroll
+        for (int t = 0; t < NF; ++t) {
+            const int f = lane + 32 * t;
+            if (f < nq) {
+                if (BF16) {
+                    const uint2 wv = reinterpret_cast<const uint2 *>(slot)[f];
+                    acc[4 * t + 0] += __uint_as_float(wv.x << 16);
+                    acc[4 * t + 1] += __uint_as_float(wv.x & 0xffff0000u);
+                    acc[4 * t + 2] += __uint_as_float(wv.y << 16);
+                    acc[4 * t + 3] += __uint_as_float(wv.y & 0xffff0000u);
+                } else {
+                    const float4 v = reinterpret_cast<const float4 *>(slot)[f];
+                    acc[4 * t + 0] += v.x;
+                    acc[4 * t + 1] += v.y;
+                    acc[4 * t + 2] += v.z;
+                    acc[4 * t + 3] += v.w;
+                }
+            }
+        }
+    }
+    __device__ __forceinline__ void finish(int lane) { flush(cur, lane); }
+};
+
+template <bool BF16, typename ACC, int NF>
+__global__ void __launch_bounds__(RS_THREADS) ring_sum_float_kernel(
+    const void *__restrict__ X, int d, const int32_t *__restrict__ perm,
+    const int32_t *__restrict__ scl, const int64_t *__restrict__ offsets, int k, ACC *__restrict__ S,
+    int64_t stride, RingLayout L, int32_t *flag) {
+    const int64_t nval = offsets[k];
+    if ((int64_t)blockIdx.x * RS_CW * RS_ROWS >= nval) return;
+    FloatCons<BF16, ACC, NF> cons;
+    cons.scl = scl;
+    cons.S = S;
+    cons.stride = stride;
+    cons.d = d;
+    ring_run(static_cast<const uint8_t *>(X), (uint32_t)d * (BF16 ? 2u : 4u), perm, nval, L, flag, cons);
+}
+
+// ------------------------------------------------------------- 1-bit rows
+// T[c][i] += Fq for every member with bit i set; T[c][d] += Fq (= U).
+// Lane l holds dimension l of every code word (t < WM words).
+template <int WM>
+struct Rbq1Cons {
+    const int32_t *scl;
+    const int64_t *fqs;  // Fq in sorted order
+    unsigned long long *T;
+    int d, W;
+    int64_t acc[WM];
+    int64_t usum;
+    int cur;
+    int64_t q0;
+    int clw, cln;
+    int64_t fqw, fqn;
+    int cnt;
+    __device__ __forceinline__ void flush(int c, int lane) {
+#pragma unroll
+        for (int t = 0; t < WM; ++t) {
+            const int col = 32 * t + lane;
+            if (t < W && col < d && acc[t])
+                atomicAdd(T + (int64_t)c * (d + 1) + col, (unsigned long long)acc[t]);
+            acc[t] = 0;
+        }
+        if (lane == 0 && usum) atomicAdd(T + (int64_t)c * (d + 1) + d, (unsigned long long)usum);
+        usum = 0;
+    }
+    __device__ __forceinline__ void start(int64_t q0_, int cnt_, int lane) {
+        q0 = q0_;
+        cnt = cnt_;
+#pragma unroll
+        for (int t = 0; t < WM; ++t) acc[t] = 0;
+        usum = 0;
+        clw = lane < cnt ? __ldg(scl + q0 + lane) : -1;
+        cln = 32 + lane < cnt ? __ldg(scl + q0 + 32 + lane) : -1;
+        fqw = lane < cnt ? __ldg(fqs + q0 + lane) : 0;
+        fqn = 32 + lane < cnt ? __ldg(fqs + q0 + 32 + lane) : 0;
+        cur = __shfl_sync(0xffffffffu, clw, 0);
+    }
+    __device__ __forceinline__ void row(int i, const uint8_t *slot, int lane) {
+        if ((i & 31) == 0 && i > 0) {
+            clw = cln;
+            fqw = fqn;
+            const int nx = i + 32 + lane;
+            cln = nx < cnt ? __ldg(scl + q0 + nx) : -1;
+            fqn = nx < cnt ? __ldg(fqs + q0 + nx) : 0;
+        }
+        const int c = __shfl_sync(0xffffffffu, clw, i & 31);
+        const int64_t fq = __shfl_sync(0xffffffffu, fqw, i & 31);
+        if (c != cur) {
+            flush(cur, lane);
+            cur = c;
+        }
+        usum += fq;
+        const uint4 *w4 = reinterpret_cast<const uint4 *>(slot);
+#pragma unroll
+        for (int g = 0; g < WM / 4; ++g) {
+            if (4 * g < W) {
+                const uint4 wv = w4[g];  // broadcast: every lane reads the same 16 bytes
+                if ((wv.x >> lane) & 1u) acc[4 * g + 0] += fq;
+                if ((wv.y >> lane) & 1u) acc[4 * g + 1] += fq;
+                if ((wv.z >> lane) & 1u) acc[4 * g + 2] += fq;
+                if ((wv.w >> lane) & 1u) acc[4 * g + 3] += fq;
+            }
+        }
+    }
+    __device__ __forceinline__ void finish(int lane) { flush(cur, lane); }
+};
+
+template <int WM>
+__global__ void __launch_bounds__(RS_THREADS) ring_sum_rbq1_kernel(
+    const uint32_t *__restrict__ codes, const int64_t *__restrict__ fqs, int d,
+    const int32_t *__restrict__ perm, const int32_t *__restrict__ scl,
+    const int64_t *__restrict__ offsets, int k, unsigned long long *__restrict__ T, RingLayout L,
+    int32_t *flag) {
+    const int64_t nval = offsets[k];
+    if ((int64_t)blockIdx.x * RS_CW * RS_ROWS >= nval) return;
+    Rbq1Cons<WM> cons;
+    cons.scl = scl;
+    cons.fqs = fqs;
+    cons.T = T;
+    cons.d = d;
+    cons.W = (d + 31) >> 5;
+    ring_run(reinterpret_cast<const uint8_t *>(codes), (uint32_t)cons.W * 4u, perm, nval, L, flag, cons);
+}
+
+bool ring_layout(uint32_t rb, RingLayout &L) {
+    if (rb == 0 || rb % 16 != 0) return false;
+    L.sb = (int)rb;
+    L.ns = (int)std::min<size_t>(RS_MAX_SLOTS, RS_RING_BYTES / ((size_t)RS_CW * rb));
+    return L.ns >= 2;
+}
+
+unsigned ring_blocks(int64_t n) {
+    const int64_t per = (int64_t)RS_CW * RS_ROWS;
+    const int64_t b = (n + per - 1) / per;
+    return (unsigned)(b < 1 ? 1 : b);
+}
+
+template <bool BF16, typename ACC>
+cudaError_t launch_float_nf(int nf, const void *X, int64_t n, int d, const int32_t *perm,
+                            const int32_t *scl, const int64_t *offsets, int k, ACC *S, RingLayout L,
+                            int32_t *flag, cudaStream_t st) {
+    const size_t smem = L.bytes();
+    const unsigned g = ring_blocks(n);
+#define RS_CASE(NFV)                                                                                \
+    case NFV: {                                                                                     \
+        auto kern = ring_sum_float_kernel<BF16, ACC, NFV>;                                          \
+        cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem); \
+        if (e != cudaSuccess) return e;                                                             \
+        kern<<<g, RS_THREADS, smem, st>>>(X, d, perm, scl, offsets, k, S, d, L, flag);               \
+        return launched();                                                                          \
+    }
+    switch (nf) {
+        RS_CASE(2)
+        RS_CASE(4)
+        RS_CASE(6)
+        RS_CASE(8)
+        RS_CASE(12)
+    default:
+        return cudaErrorInvalidValue;
+    }
+#undef RS_CASE
+}
+
+}  // namespace
+
+bool ring_sum_float_ok(const void *X, int x_is_bf16, int d) {
+    RingLayout L;
+    const uint32_t rb = (uint32_t)d * (x_is_bf16 ? 2u : 4u);
+    return d % 4 == 0 && (reinterpret_cast<uintptr_t>(X) & 15u) == 0 && d <= 12 * 128 &&
+           ring_layout(rb, L);
+}
+
+bool ring_sum_rbq1_ok(const void *codes, int d) {
+    RingLayout L;
+    const int W = (d + 31) >> 5;
+    return W % 4 == 0 && W <= 32 && (reinterpret_cast<uintptr_t>(codes) & 15u) == 0 &&
+           ring_layout((uint32_t)W * 4u, L);
+}
+
+cudaError_t launch_ring_sum_float(const void *X, int x_is_bf16, int64_t n, int d, const int32_t *perm,
+                                  const int32_t *scl, const int64_t *offsets, int k, float *S_f,
+                                  double *S_d, int32_t *flag, cudaStream_t st) {
+    if (n == 0) return cudaSuccess;
+    RingLayout L;
+    if (!ring_layout((uint32_t)d * (x_is_bf16 ? 2u : 4u), L)) return cudaErrorInvalidValue;
+    const int q = (d / 4 + 31) / 32;  // float4 groups per lane
+    const int nf = q <= 2 ? 2 : q <= 4 ? 4 : q <= 6 ? 6 : q <= 8 ? 8 : 12;
+    if (S_d)
+        return x_is_bf16 ? launch_float_nf<true, double>(nf, X, n, d, perm, scl, offsets, k, S_d, L, flag, st)
+                         : launch_float_nf<false, double>(nf, X, n, d, perm, scl, offsets, k, S_d, L, flag, st);
+    return x_is_bf16 ? launch_float_nf<true, float>(nf, X, n, d, perm, scl, offsets, k, S_f, L, flag, st)
+                     : launch_float_nf<false, float>(nf, X, n, d, perm, scl, offsets, k, S_f, L, flag, st);
+}
+
+cudaError_t launch_ring_sum_rbq1(const uint32_t *codes, const int64_t *fqs, int64_t n, int d,
+                                 const int32_t *perm, const int32_t *scl, const int64_t *offsets,
+                                 int k, int64_t *T, int32_t *flag, cudaStream_t st) {
+    if (n == 0) return cudaSuccess;
+    const int W = (d + 31) >> 5;
+    RingLayout L;
+    if (!ring_layout((uint32_t)W * 4u, L)) return cudaErrorInvalidValue;
+    const size_t smem = L.bytes();
+    const unsigned g = ring_blocks(n);
+    auto T64 = reinterpret_cast<unsigned long long *>(T);
+#define RS_CASE(WMV)                                                                                \
+    if (W <= WMV) {                                                                                 \
+        auto kern = ring_sum_rbq1_kernel<WMV>;                                                      \
+        cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem); \
+        if (e != cudaSuccess) return e;                                                             \
+        kern<<<g, RS_THREADS, smem, st>>>(codes, fqs, d, perm, scl, offsets, k, T64, L, flag);       \
+        return launched();                                                                          \
+    }
+    RS_CASE(8)
+    RS_CASE(16)
+    RS_CASE(24)
+    RS_CASE(32)
+#undef RS_CASE
+    return cudaErrorInvalidValue;
+}
+
+}  // namespace skm

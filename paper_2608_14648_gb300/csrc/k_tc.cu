@@ -6,11 +6,12 @@
 //               (bf16, 128-byte swizzle) per stage, 4-stage mbarrier ring
 //   warp 1      MMA issuer: 4 x tcgen05.mma.kind::f16 (M=128, N=256, K=16)
 //               per stage into one of two 128 x 256 fp32 TMEM accumulators
-//   warps 2-9   epilogue: tcgen05.ld of the accumulator (thread = point row;
-//               two warps per TMEM lane quarter, each taking half of the 256
+//   warps 2..   epilogue: tcgen05.ld of the accumulator (thread = point row;
+//               NH warps per TMEM lane quarter, each taking 256 / NH of the
 //               columns), fused per-row reduction over centroids, so the
-//               N x K distance matrix never leaves the SM; the two halves of a
-//               row merge through shared memory at the end of a point tile
+//               N x K distance matrix never leaves the SM; the NH column
+//               slices of a row merge through shared memory at the end of a
+//               point tile
 // Two epilogues:
 //  SCREEN (fp32 / bf16 points): bf16 operands, so the dot product carries a
 //    rounding error.  Each pair gets a rigorous interval [L, U] for
@@ -48,15 +49,28 @@ constexpr int BK = 64;   // bf16 elements per 128-byte swizzle row
 constexpr int STAGES = 4;
 constexpr int A_STAGE = BM * BK * 2;  // 16 KiB
 constexpr int B_STAGE = BN * BK * 2;  // 32 KiB
-constexpr int EPI_WARPS = 8;  // two per TMEM lane quarter
-constexpr int THREADS = 64 + 32 * EPI_WARPS;
 constexpr int TCAND = 4;
 constexpr unsigned long long WAIT_LIMIT_NS = 2000000000ull;  // 2 s per barrier wait
-constexpr int MERGE_WORDS = 2 * TCAND + 2;                    // one row's screen state
-constexpr int MERGE_BYTES = 2 * BM * MERGE_WORDS * 4;         // double-buffered by point tile
-constexpr size_t SMEM_BYTES = 1024 + (size_t)STAGES * (A_STAGE + B_STAGE) + 256 + MERGE_BYTES;
 
 enum { MODE_SCREEN = 0, MODE_SQ8 = 1, MODE_RBQ1 = 2 };
+// epilogue warps per TMEM lane quarter, by mode
+constexpr int TC_NH[3] = {4, 2, 4};
+
+// Epilogue shape: NH warps per TMEM lane quarter (column slices of 256 / NH).
+template <int NH>
+constexpr int epi_threads() { return 128 * NH; }
+template <int NH>
+constexpr int tc_threads() { return 64 + epi_threads<NH>(); }
+// one row's state for the merge: the screen list, or (best, index)
+template <int MODE>
+constexpr int merge_words() { return MODE == MODE_SCREEN ? 2 * TCAND + 2 : 2; }
+// 1024-byte alignment slack, the stages, barriers + TMEM slot (352 bytes), and
+// the merge buffer: slices 1..NH-1 publish, double-buffered by point tile
+template <int MODE, int NH>
+constexpr size_t tc_smem_bytes() {
+    return 1024 + (size_t)STAGES * (A_STAGE + B_STAGE) + 512 +
+           (size_t)2 * (NH - 1) * BM * merge_words<MODE>() * 4;
+}
 
 struct TcParams {
     int64_t n;
@@ -295,8 +309,8 @@ __device__ __forceinline__ void screen_insert(ScreenRow &s, float L, int j) {
     }
 }
 
-template <int MODE>
-__global__ void __launch_bounds__(THREADS, 1)
+template <int MODE, int NH>
+__global__ void __launch_bounds__(tc_threads<NH>(), 1)
     tc_assign_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                      const TcParams p) {
     extern __shared__ uint8_t smem_raw[];
@@ -312,7 +326,7 @@ __global__ void __launch_bounds__(THREADS, 1)
     auto tfull_bar = [&](int b) { return bar0 + 8u * (2 * STAGES + b); };
     auto tempty_bar = [&](int b) { return bar0 + 8u * (2 * STAGES + 2 + b); };
     uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(bars + 2 * STAGES + 4);
-    // the epilogue's merge buffer starts 256 bytes after tmem_slot (see SMEM_BYTES)
+    // the epilogue's merge buffer starts 256 bytes after tmem_slot (see tc_smem_bytes)
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     volatile int32_t *abort_flag = p.counters + 2;
@@ -325,7 +339,7 @@ __global__ void __launch_bounds__(THREADS, 1)
         }
         for (int b = 0; b < 2; ++b) {
             mbar_init(tfull_bar(b), 1);
-            mbar_init(tempty_bar(b), EPI_WARPS * 32);
+            mbar_init(tempty_bar(b), epi_threads<NH>());
         }
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
         asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmA)) : "memory");
@@ -386,11 +400,13 @@ __global__ void __launch_bounds__(THREADS, 1)
         mma_done:;
         }
     } else {  // ------------------------------------------------------- epilogue
-        const int e = warp - 2;          // 0..7
+        constexpr int SW = BN / NH;      // columns per slice
+        constexpr int MW = merge_words<MODE>();
+        const int e = warp - 2;          // 0 .. 4 NH - 1
         const int q = warp & 3;          // TMEM lane quarter this warp may access
-        const int half = e >> 2;         // which 128 of the 256 columns
+        const int slice = e >> 2;        // which SW of the 256 columns
         const int rin = q * 32 + lane;   // row within the point tile
-        uint32_t *merge = reinterpret_cast<uint32_t *>(tmem_slot + 64);  // [2][BM][MERGE_WORDS]
+        uint32_t *merge = reinterpret_cast<uint32_t *>(tmem_slot + 64);  // [2][NH-1][BM][MW]
         uint32_t job = 0;
         uint32_t tile = 0;
         for (int64_t rt = blockIdx.x; rt < p.nrt; rt += gridDim.x, ++tile) {
@@ -416,10 +432,10 @@ __global__ void __launch_bounds__(THREADS, 1)
                 const bool ok = mbar_wait(tfull_bar(b), bph, abort_flag);
                 if (!__all_sync(0xffffffffu, ok)) goto epi_done;
                 tc_fence_after();
-                const uint32_t taddr = tmem + ((uint32_t)(q * 32) << 16) + b * BN + half * (BN / 2);
-                const int jh = ct * BN + half * (BN / 2);
+                const uint32_t taddr = tmem + ((uint32_t)(q * 32) << 16) + b * BN + slice * SW;
+                const int jh = ct * BN + slice * SW;
 #pragma unroll 1
-                for (int c = 0; c < BN / 64; ++c) {
+                for (int c = 0; c < SW / 32; ++c) {
                     const int j0 = jh + c * 32;
                     if (j0 >= p.k) break;  // warp-uniform
                     uint32_t v[32];
@@ -478,7 +494,8 @@ __global__ void __launch_bounds__(THREADS, 1)
                         // fp32 order (u = fma(sd, 2P - sum ybar, bd pc),
                         // est = fma(-2F, u, nx2 + ny2)).  The e4m3
                         // accumulator carries a small non-integer error (~2^-12),
-                        // so P is its nearest integer; 2P - sum ybar is exact.
+                        // so P is its nearest integer, taken as (acc + 2^23) - 2^23
+                        // (exact for 0 <= acc < 2^22); 2P - sum ybar is exact.
                         float gb[4];
                         int gi[4];
 #pragma unroll
@@ -492,8 +509,10 @@ __global__ void __launch_bounds__(THREADS, 1)
                                 const float4 qn = __ldg(p.rinfoq + ((j0 + i) >> 1));
                                 // packed pairs; every product here feeds an explicit fma
                                 // (no separate multiply-add the compiler could fuse)
-                                const float2 P2 = make_float2(rintf(__uint_as_float(v[i])),
-                                                              rintf(__uint_as_float(v[i + 1])));
+                                const float2 P2 = fsub2(
+                                    fadd2(make_float2(__uint_as_float(v[i]), __uint_as_float(v[i + 1])),
+                                          make_float2(0x1p23f, 0x1p23f)),
+                                    make_float2(0x1p23f, 0x1p23f));
                                 const float2 qv = ffma2(make_float2(2.0f, 2.0f), P2, make_float2(qn.x, qn.y));
                                 const float2 t = fmul2(make_float2(bs.x, bs.y), make_float2(rpc, rpc));
                                 const float2 u = ffma2(make_float2(bs.z, bs.w), qv, t);
@@ -521,9 +540,9 @@ __global__ void __launch_bounds__(THREADS, 1)
                 tc_fence_before();
                 mbar_arrive(tempty_bar(b));
             }
-            // merge the two column halves of each row: half 1 publishes, half 0 finishes
-            uint32_t *slot = merge + ((tile & 1u) * BM + rin) * MERGE_WORDS;
-            if (half == 1) {
+            // merge the column slices of each row: slices 1.. publish, slice 0 finishes
+            if (slice > 0) {
+                uint32_t *slot = merge + (((tile & 1u) * (NH - 1) + (slice - 1)) * BM + rin) * MW;
                 if (MODE == MODE_SCREEN) {
 #pragma unroll
                     for (int t = 0; t < TCAND; ++t) {
@@ -540,14 +559,34 @@ __global__ void __launch_bounds__(THREADS, 1)
                     slot[1] = (uint32_t)besti;
                 }
             }
-            asm volatile("bar.sync 1, %0;" ::"n"(EPI_WARPS * 32) : "memory");
-            if (half == 0 && valid) {
-                if (MODE == MODE_SCREEN) {
-                    sr.umin = fminf(sr.umin, __uint_as_float(slot[2 * TCAND]));
-                    sr.lev = fminf(sr.lev, __uint_as_float(slot[2 * TCAND + 1]));
+            asm volatile("bar.sync 1, %0;" ::"n"(epi_threads<NH>()) : "memory");
+            if (slice == 0 && valid) {
+                // slices in increasing column order; ties resolve to the lower index
 #pragma unroll
-                    for (int t = 0; t < TCAND; ++t)
-                        screen_insert(sr, __uint_as_float(slot[t]), (int)slot[TCAND + t]);
+                for (int h = 1; h < NH; ++h) {
+                    const uint32_t *slot = merge + (((tile & 1u) * (NH - 1) + (h - 1)) * BM + rin) * MW;
+                    if (MODE == MODE_SCREEN) {
+                        sr.umin = fminf(sr.umin, __uint_as_float(slot[2 * TCAND]));
+                        sr.lev = fminf(sr.lev, __uint_as_float(slot[2 * TCAND + 1]));
+#pragma unroll
+                        for (int t = 0; t < TCAND; ++t)
+                            screen_insert(sr, __uint_as_float(slot[t]), (int)slot[TCAND + t]);
+                    } else if (MODE == MODE_SQ8) {
+                        const int32_t ob = (int32_t)slot[0], oi = (int32_t)slot[1];
+                        if (ob < best || (ob == best && oi < besti)) {
+                            best = ob;
+                            besti = oi;
+                        }
+                    } else {
+                        const float ob = __uint_as_float(slot[0]);
+                        const int32_t oi = (int32_t)slot[1];
+                        if (ob < fbest || (ob == fbest && oi < besti)) {
+                            fbest = ob;
+                            besti = oi;
+                        }
+                    }
+                }
+                if (MODE == MODE_SCREEN) {
                     int ncert = 0;
 #pragma unroll
                     for (int t = 0; t < TCAND; ++t) ncert += (sr.L[t] <= sr.umin) ? 1 : 0;
@@ -566,20 +605,9 @@ __global__ void __launch_bounds__(THREADS, 1)
                         p.fall_rows[atomicAdd(&p.counters[1], 1)] = (int32_t)row;
                     }
                 } else if (MODE == MODE_SQ8) {
-                    const int32_t ob = (int32_t)slot[0], oi = (int32_t)slot[1];
-                    if (ob < best || (ob == best && oi < besti)) {
-                        best = ob;
-                        besti = oi;
-                    }
                     p.assign[row] = besti;
                     if (p.dist) p.dist[row] = (float)best;
                 } else {
-                    const float ob = __uint_as_float(slot[0]);
-                    const int32_t oi = (int32_t)slot[1];
-                    if (ob < fbest || (ob == fbest && oi < besti)) {
-                        fbest = ob;
-                        besti = oi;
-                    }
                     p.assign[row] = besti;
                     if (p.dist) p.dist[row] = fbest;
                 }
@@ -921,12 +949,14 @@ int device_sms() {
 template <int MODE>
 int launch_tc(const void *xs, int64_t n, int dp, int d, const void *cs, int k, const TcParams &p0,
               cudaStream_t st) {
+    constexpr int NH = TC_NH[MODE];
+    constexpr size_t SMEM = tc_smem_bytes<MODE, NH>();
+    static_assert(SMEM <= 227 * 1024, "shared memory per CTA");
     static std::once_flag attr_once[3];
     static cudaError_t attr_err[3] = {cudaSuccess, cudaSuccess, cudaSuccess};
     std::call_once(attr_once[MODE], [] {
-        attr_err[MODE] = cudaFuncSetAttribute(tc_assign_kernel<MODE>,
-                                              cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                              (int)SMEM_BYTES);
+        attr_err[MODE] = cudaFuncSetAttribute(tc_assign_kernel<MODE, NH>,
+                                              cudaFuncAttributeMaxDynamicSharedMemorySize, (int)SMEM);
     });
     if (attr_err[MODE] != cudaSuccess)
         return set_error(SKM_ERR_CUDA, "cudaFuncSetAttribute: %s", cudaGetErrorString(attr_err[MODE]));
@@ -941,7 +971,7 @@ int launch_tc(const void *xs, int64_t n, int dp, int d, const void *cs, int k, c
     p.nct = (int)cdiv(k, BN);
     p.nkc = (int)cdiv(d, 128 / eb);
     const int grid = (int)std::min<int64_t>(device_sms(), p.nrt);
-    tc_assign_kernel<MODE><<<grid, THREADS, SMEM_BYTES, st>>>(ma, mb, p);
+    tc_assign_kernel<MODE, NH><<<grid, tc_threads<NH>(), SMEM, st>>>(ma, mb, p);
     SKM_CUDA_TRY(launched());
     return SKM_OK;
 }

@@ -107,9 +107,50 @@ __global__ void scatter_kernel(const int32_t *__restrict__ assign, int64_t n, in
     }
 }
 
+// Block-aggregated form: a block counts its SC_POINTS points per cluster in
+// shared memory, reserves one range per cluster with a single global atomic,
+// then places its points inside those ranges (shared-memory atomics), so the
+// global atomics drop from one per point to one per (block, cluster).
+constexpr int SC_POINTS = 4096;
+constexpr int SC_THREADS = 512;
+constexpr int SC_MAX_K = 12288;  // 48 KiB of counters
+
+__global__ void __launch_bounds__(SC_THREADS) scatter_blocked_kernel(
+    const int32_t *__restrict__ assign, int64_t n, int k, const int64_t *__restrict__ offsets,
+    int32_t *__restrict__ cursor, int32_t *__restrict__ perm, int32_t *__restrict__ scl) {
+    extern __shared__ int32_t cnt_sh[];
+    const int64_t p0 = (int64_t)blockIdx.x * SC_POINTS;
+    const int64_t p1 = min(n, p0 + SC_POINTS);
+    for (int j = threadIdx.x; j < k; j += SC_THREADS) cnt_sh[j] = 0;
+    __syncthreads();
+    for (int64_t t = p0 + threadIdx.x; t < p1; t += SC_THREADS) {
+        const int a = assign[t];
+        if (a >= 0 && a < k) atomicAdd(&cnt_sh[a], 1);
+    }
+    __syncthreads();
+    for (int j = threadIdx.x; j < k; j += SC_THREADS) {
+        const int c = cnt_sh[j];
+        if (c) cnt_sh[j] = (int32_t)offsets[j] + atomicAdd(&cursor[j], c);
+    }
+    __syncthreads();
+    for (int64_t t = p0 + threadIdx.x; t < p1; t += SC_THREADS) {
+        const int a = assign[t];
+        if (a < 0 || a >= k) continue;  // skipped consistently with the histogram
+        const int pos = atomicAdd(&cnt_sh[a], 1);
+        perm[pos] = (int32_t)t;
+        if (scl) scl[pos] = a;
+    }
+}
+
 cudaError_t launch_scatter(const int32_t *assign, int64_t n, int k, const int64_t *offsets,
                            int32_t *cursor, int32_t *perm, int32_t *scl, cudaStream_t st) {
     if (n == 0) return cudaSuccess;
+    if (k <= SC_MAX_K) {
+        const int64_t blocks = (n + SC_POINTS - 1) / SC_POINTS;
+        scatter_blocked_kernel<<<(unsigned)blocks, SC_THREADS, sizeof(int32_t) * (size_t)k, st>>>(
+            assign, n, k, offsets, cursor, perm, scl);
+        return launched();
+    }
     int64_t blocks = (n + 255) / 256;
     if (blocks > 152 * 8) blocks = 152 * 8;
     scatter_kernel<<<(unsigned)blocks, 256, 0, st>>>(assign, n, k, offsets, cursor, perm, scl);
@@ -247,20 +288,24 @@ __device__ __forceinline__ float rbq1_finish(int64_t T, int64_t U, int64_t cnt, 
     return __double2float_rn(__dadd_rn((double)m, v));
 }
 
-// Fixed-point weights Fq = rint(F 2^e), once per update call.
-__global__ void rbq1_fq_kernel(const float *__restrict__ F, int64_t n, int e,
+// Fixed-point weights Fq = rint(F 2^e), once per update call, written in the
+// cluster-sorted order (position q holds the weight of member perm[q]).
+__global__ void rbq1_fq_kernel(const float *__restrict__ F, const int32_t *__restrict__ perm,
+                               const int64_t *__restrict__ offsets, int k, int e,
                                int64_t *__restrict__ fq) {
     const double pow2 = ldexp(1.0, e);
-    for (int64_t t = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; t < n;
-         t += (int64_t)gridDim.x * blockDim.x)
-        fq[t] = __double2ll_rn(__dmul_rn((double)F[t], pow2));
+    const int64_t nval = offsets[k];
+    for (int64_t q = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; q < nval;
+         q += (int64_t)gridDim.x * blockDim.x)
+        fq[q] = __double2ll_rn(__dmul_rn((double)F[perm[q]], pow2));
 }
 
-cudaError_t launch_rbq1_fq(const float *F, int64_t n, int e, int64_t *fq, cudaStream_t st) {
+cudaError_t launch_rbq1_fq(const float *F, const int32_t *perm, const int64_t *offsets, int k,
+                           int64_t n, int e, int64_t *fq, cudaStream_t st) {
     int64_t blocks = (n + 255) / 256;
     if (blocks > 152 * 8) blocks = 152 * 8;
     if (blocks < 1) blocks = 1;
-    rbq1_fq_kernel<<<(int)blocks, 256, 0, st>>>(F, n, e, fq);
+    rbq1_fq_kernel<<<(int)blocks, 256, 0, st>>>(F, perm, offsets, k, e, fq);
     return launched();
 }
 
@@ -335,7 +380,8 @@ __global__ void __launch_bounds__(CH_WARPS * 32) chunk_sum_float_kernel(
     }
 }
 
-// 1-bit codes -> int64 accumulators T[k][d+1] (column d holds U = sum Fq).
+// 1-bit codes -> int64 accumulators T[k][d+1] (column d holds U = sum Fq);
+// fqs in the sorted order.
 __global__ void __launch_bounds__(CH_WARPS * 32) chunk_sum_rbq1_kernel(
     const uint32_t *__restrict__ codes, const int64_t *__restrict__ fqs, int d,
     const int32_t *__restrict__ perm, const int32_t *__restrict__ scl,
@@ -367,7 +413,7 @@ __global__ void __launch_bounds__(CH_WARPS * 32) chunk_sum_rbq1_kernel(
         for (int64_t q = q0; q < q1; ++q) {
             const int c = scl[q];
             const int64_t p = perm[q];
-            const int64_t fq = __ldg(fqs + p);
+            const int64_t fq = __ldg(fqs + q);
             const uint32_t mine = (lane < nw) ? __ldg(codes + p * W + w0 + lane) : 0u;
             if (c != cur) {
                 flush(cur);

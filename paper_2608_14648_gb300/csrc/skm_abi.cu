@@ -118,6 +118,7 @@ struct UpdateBufs {
     int64_t *fq = nullptr;    // RBQ1: fixed-point weights round(F 2^e)
     float *sumf = nullptr;    // F32/BF16: cluster sums [k][d]
     int64_t *sumi = nullptr;  // RBQ1: cluster sums [k][d + 1]
+    int32_t *flag = nullptr;  // raised by a streamed-sum wait that gave up
 };
 
 static void plan_update(const skm_data *x, int k, Carver &cv, UpdateBufs &b) {
@@ -131,6 +132,7 @@ static void plan_update(const skm_data *x, int k, Carver &cv, UpdateBufs &b) {
         b.sumi = cv.take<int64_t>((size_t)k * (x->d + 1));
     }
     if (x->repr == SKM_REPR_F32 || x->repr == SKM_REPR_BF16) b.sumf = cv.take<float>((size_t)k * x->d);
+    b.flag = cv.take<int32_t>(1);
 }
 
 struct FitBufs {
@@ -222,29 +224,36 @@ static int do_update(const skm_data *x, const int32_t *assign, int k, void *C, i
     SKM_CUDA_TRY(launch_scatter(assign, n, k, b.offsets, b.cursor, b.perm, b.scl, st));
     switch (x->repr) {
     case SKM_REPR_F32:
-    case SKM_REPR_BF16:
-        if (partial) {
-            SKM_CUDA_TRY(launch_chunk_sum_float(x->x, x->repr == SKM_REPR_BF16, n, d, b.perm, b.scl,
-                                                b.offsets, k, nullptr,
-                                                static_cast<double *>(partial), st));
-        } else {
-            SKM_CUDA_TRY(cudaMemsetAsync(b.sumf, 0, sizeof(float) * (size_t)k * d, st));
-            SKM_CUDA_TRY(launch_chunk_sum_float(x->x, x->repr == SKM_REPR_BF16, n, d, b.perm, b.scl,
-                                                b.offsets, k, b.sumf, nullptr, st));
+    case SKM_REPR_BF16: {
+        const int bf = x->repr == SKM_REPR_BF16;
+        const bool ring = ring_sum_float_ok(x->x, bf, d);
+        float *Sf = partial ? nullptr : b.sumf;
+        double *Sd = partial ? static_cast<double *>(partial) : nullptr;
+        if (!partial) SKM_CUDA_TRY(cudaMemsetAsync(b.sumf, 0, sizeof(float) * (size_t)k * d, st));
+        if (ring)
+            SKM_CUDA_TRY(launch_ring_sum_float(x->x, bf, n, d, b.perm, b.scl, b.offsets, k, Sf, Sd,
+                                               b.flag, st));
+        else
+            SKM_CUDA_TRY(launch_chunk_sum_float(x->x, bf, n, d, b.perm, b.scl, b.offsets, k, Sf, Sd, st));
+        if (!partial)
             SKM_CUDA_TRY(launch_finalize_float32(b.sumf, counts, k, d, static_cast<float *>(C), st));
-        }
         break;
+    }
     case SKM_REPR_SQ8:
         SKM_CUDA_TRY(launch_segsum_sq8(static_cast<const uint8_t *>(x->x), d, b.perm, b.offsets, k,
                                        static_cast<uint8_t *>(C), static_cast<int64_t *>(partial),
                                        st));
         break;
     case SKM_REPR_RBQ1: {
-        SKM_CUDA_TRY(launch_rbq1_fq(x->F, n, e, b.fq, st));
+        SKM_CUDA_TRY(launch_rbq1_fq(x->F, b.perm, b.offsets, k, n, e, b.fq, st));
         int64_t *T = partial ? static_cast<int64_t *>(partial) : b.sumi;
         if (!partial) SKM_CUDA_TRY(cudaMemsetAsync(T, 0, sizeof(int64_t) * (size_t)k * (d + 1), st));
-        SKM_CUDA_TRY(launch_chunk_sum_rbq1(static_cast<const uint32_t *>(x->x), b.fq, n, d, b.perm,
-                                           b.scl, b.offsets, k, T, st));
+        const uint32_t *codes = static_cast<const uint32_t *>(x->x);
+        if (ring_sum_rbq1_ok(codes, d))
+            SKM_CUDA_TRY(launch_ring_sum_rbq1(codes, b.fq, n, d, b.perm, b.scl, b.offsets, k, T,
+                                              b.flag, st));
+        else
+            SKM_CUDA_TRY(launch_chunk_sum_rbq1(codes, b.fq, n, d, b.perm, b.scl, b.offsets, k, T, st));
         if (!partial)
             SKM_CUDA_TRY(launch_finalize_rbq1(T, counts, k, d, x->m, e, static_cast<float *>(C), st));
         break;
@@ -478,6 +487,7 @@ int skm_update(const skm_data *x, const int32_t *assign, int k, void *C_inout, i
     UpdateBufs b;
     plan_update(x, k, cv, b);
     SKM_TRY(need_ws(cv, ws_bytes, ws));
+    SKM_CUDA_TRY(cudaMemsetAsync(b.flag, 0, sizeof(int32_t), S(stream)));
     return do_update(x, assign, k, C_inout, counts, partial, x->rbq1_exp, b, S(stream));
 }
 
@@ -550,6 +560,7 @@ int skm_fit(const skm_fit_config *cfg, const skm_data *x, const void *C_init,
     }
     // STEP 1: initial centroids
     SKM_CUDA_TRY(cudaMemsetAsync(b.status, 0, sizeof(int), st));
+    SKM_CUDA_TRY(cudaMemsetAsync(b.u.flag, 0, sizeof(int32_t), st));
     if (C_init) {
         SKM_CUDA_TRY(cudaMemcpyAsync(C_out, C_init, centroid_bytes(x, k), cudaMemcpyDeviceToDevice,
                                      st));
@@ -589,6 +600,9 @@ int skm_fit(const skm_fit_config *cfg, const skm_data *x, const void *C_init,
     skm_stats local;
     memset(&local, 0, sizeof(local));
     SKM_TRY(tc_read_stats(b.a.tc, &local, st));
+    int32_t uflag = 0;
+    SKM_CUDA_TRY(cudaMemcpy(&uflag, b.u.flag, sizeof(uflag), cudaMemcpyDeviceToHost));
+    if (uflag) return set_error(SKM_ERR_TIMEOUT, "an update pipeline wait exceeded its limit");
     unsigned long long pr[2] = {0, 0};
     SKM_CUDA_TRY(cudaMemcpy(pr, b.a.prune, sizeof(pr), cudaMemcpyDeviceToHost));
     local.prune_first_block = (int64_t)pr[0];

@@ -123,7 +123,7 @@ cudaError_t launch_chunk_sum_float(const void *X, int x_is_bf16, int64_t n, int 
                                    const int32_t *perm, const int32_t *scl,
                                    const int64_t *offsets, int k, float *S_f, double *S_d,
                                    cudaStream_t st);
-cudaError_t launch_chunk_sum_rbq1(const uint32_t *codes, const int64_t *fq, int64_t n, int d,
+cudaError_t launch_chunk_sum_rbq1(const uint32_t *codes, const int64_t *fq_sorted, int64_t n, int d,
                                   const int32_t *perm, const int32_t *scl, const int64_t *offsets,
                                   int k, int64_t *T, cudaStream_t st);
 cudaError_t launch_finalize_float32(const float *S, const int64_t *counts, int k, int d,
@@ -131,7 +131,19 @@ cudaError_t launch_finalize_float32(const float *S, const int64_t *counts, int k
 cudaError_t launch_segsum_sq8(const uint8_t *X, int d, const int32_t *perm,
                               const int64_t *offsets, int k, uint8_t *C_inout, int64_t *partial,
                               cudaStream_t st);
-cudaError_t launch_rbq1_fq(const float *F, int64_t n, int e, int64_t *fq, cudaStream_t st);
+// Fq = round(F[perm[q]] 2^e) for the sorted positions q < offsets[k]
+cudaError_t launch_rbq1_fq(const float *F, const int32_t *perm, const int64_t *offsets, int k,
+                           int64_t n, int e, int64_t *fq_sorted, cudaStream_t st);
+// streamed segmented sums (cp.async.bulk row gathers into shared-memory rings);
+// *_ok says whether the row size and alignment suit them
+bool ring_sum_float_ok(const void *X, int x_is_bf16, int d);
+bool ring_sum_rbq1_ok(const void *codes, int d);
+cudaError_t launch_ring_sum_float(const void *X, int x_is_bf16, int64_t n, int d, const int32_t *perm,
+                                  const int32_t *scl, const int64_t *offsets, int k, float *S_f,
+                                  double *S_d, int32_t *flag, cudaStream_t st);
+cudaError_t launch_ring_sum_rbq1(const uint32_t *codes, const int64_t *fq_sorted, int64_t n, int d,
+                                 const int32_t *perm, const int32_t *scl, const int64_t *offsets,
+                                 int k, int64_t *T, int32_t *flag, cudaStream_t st);
 cudaError_t launch_finalize_float(const double *partial, const int64_t *counts, int k, int d,
                                   float *C_inout, cudaStream_t st);
 cudaError_t launch_finalize_sq8(const int64_t *partial, const int64_t *counts, int k, int d,
