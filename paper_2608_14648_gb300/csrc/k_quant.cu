@@ -133,15 +133,36 @@ cudaError_t launch_sq8_decode(const uint8_t *codes, int64_t n, int d, const floa
     return launched();
 }
 
+// Column sums: each block sums a contiguous run of rows; a thread owns
+// columns c, c + 256, ... and keeps a Kahan-compensated fp32 sum per column
+// (error about 2^-23 of the sum of magnitudes), written out as fp64.
 __global__ void colsum_partial_kernel(const float *__restrict__ X, int64_t n, int d,
                                       double *__restrict__ psum) {
     const int64_t rows_per = (n + gridDim.x - 1) / gridDim.x;
     const int64_t r0 = (int64_t)blockIdx.x * rows_per;
     const int64_t r1 = min(n, r0 + rows_per);
     for (int c = threadIdx.x; c < d; c += blockDim.x) {
-        double acc = 0.0;
-        for (int64_t r = r0; r < r1; ++r) acc += (double)X[r * d + c];
-        psum[(int64_t)blockIdx.x * d + c] = acc;
+        float s = 0.0f, comp = 0.0f;
+        int64_t r = r0;
+        for (; r + 4 <= r1; r += 4) {
+            float v[4];
+#pragma unroll
+            for (int u = 0; u < 4; ++u) v[u] = __ldg(X + (r + u) * d + c);
+#pragma unroll
+            for (int u = 0; u < 4; ++u) {
+                const float y = __fsub_rn(v[u], comp);
+                const float t = __fadd_rn(s, y);
+                comp = __fsub_rn(__fsub_rn(t, s), y);
+                s = t;
+            }
+        }
+        for (; r < r1; ++r) {
+            const float y = __fsub_rn(__ldg(X + r * d + c), comp);
+            const float t = __fadd_rn(s, y);
+            comp = __fsub_rn(__fsub_rn(t, s), y);
+            s = t;
+        }
+        psum[(int64_t)blockIdx.x * d + c] = (double)s - (double)comp;
     }
 }
 
@@ -171,8 +192,19 @@ cudaError_t launch_colmean_finish(const double *psum, int nblk, int d, int64_t n
 // ---------------------------------------------------------------------------
 // RabitQ 1-bit encode: one warp per point.  Lane l handles dimensions
 // 32w + l; the sign bits of a 32-dimension group are one __ballot_sync.
-// ||r||^2 and ||r||_1 are fp64 (lane partials, fixed xor-tree reduction).
+// ||r||^2 and ||r||_1: Kahan-compensated fp32 lane sums (relative error about
+// 2^-23), then an fp64 xor-tree across lanes; F = sqrt(d) ||r||^2 / ||r||_1
+// is evaluated in fp64 and rounded once.
 // ---------------------------------------------------------------------------
+__device__ __forceinline__ void kahan_add(float &s, float &c, float v) {
+    const float y = __fsub_rn(v, c);
+    const float t = __fadd_rn(s, y);
+    c = __fsub_rn(__fsub_rn(t, s), y);
+    s = t;
+}
+
+constexpr int ENC_UNROLL = 8;
+
 __global__ void rbq1_encode_kernel(const float *__restrict__ X, int64_t n, int d,
                                    const float *__restrict__ m, uint32_t *__restrict__ codes,
                                    float *__restrict__ nx2, float *__restrict__ F,
@@ -181,33 +213,43 @@ __global__ void rbq1_encode_kernel(const float *__restrict__ X, int64_t n, int d
     const int64_t warp = (blockIdx.x * (int64_t)blockDim.x + threadIdx.x) >> 5;
     const int64_t nwarps = ((int64_t)gridDim.x * blockDim.x) >> 5;
     const int W = (d + 31) >> 5;
+    const double sqrt_d = sqrt((double)d);
     for (int64_t p = warp; p < n; p += nwarps) {
         const float *x = X + p * d;
-        double s2 = 0.0, s1 = 0.0;
+        float s2 = 0.0f, c2 = 0.0f, s1 = 0.0f, c1 = 0.0f;
         int pc = 0;
-        for (int w = 0; w < W; ++w) {
-            const int i = 32 * w + lane;
-            float r = 0.0f;
-            if (i < d) r = __fsub_rn(x[i], m[i]);
-            const unsigned bits = __ballot_sync(0xffffffffu, r > 0.0f);
-            const double rd = (double)r;
-            s2 = __fma_rn(rd, rd, s2);
-            s1 = __dadd_rn(s1, fabs(rd));
-            if (lane == 0) {
-                codes[p * W + w] = bits;
-                pc += __popc(bits);
+        for (int w0 = 0; w0 < W; w0 += ENC_UNROLL) {
+            float v[ENC_UNROLL];
+#pragma unroll
+            for (int u = 0; u < ENC_UNROLL; ++u) {
+                const int i = 32 * (w0 + u) + lane;
+                v[u] = (w0 + u < W && i < d) ? __ldg(x + i) : 0.0f;
+            }
+#pragma unroll
+            for (int u = 0; u < ENC_UNROLL; ++u) {
+                const int w = w0 + u;
+                if (w < W) {  // warp-uniform
+                    const int i = 32 * w + lane;
+                    const float r = i < d ? __fsub_rn(v[u], __ldg(m + i)) : 0.0f;
+                    const unsigned bits = __ballot_sync(0xffffffffu, r > 0.0f);
+                    kahan_add(s2, c2, __fmul_rn(r, r));
+                    kahan_add(s1, c1, fabsf(r));
+                    if (lane == 0) {
+                        codes[p * W + w] = bits;
+                        pc += __popc(bits);
+                    }
+                }
             }
         }
+        double t2 = (double)s2 - (double)c2, t1 = (double)s1 - (double)c1;
 #pragma unroll
         for (int o = 16; o > 0; o >>= 1) {
-            s2 += __shfl_xor_sync(0xffffffffu, s2, o);
-            s1 += __shfl_xor_sync(0xffffffffu, s1, o);
+            t2 += __shfl_xor_sync(0xffffffffu, t2, o);
+            t1 += __shfl_xor_sync(0xffffffffu, t1, o);
         }
         if (lane == 0) {
-            nx2[p] = __double2float_rn(s2);
-            F[p] = (s1 > 0.0)
-                       ? __double2float_rn(__ddiv_rn(__dmul_rn(__dsqrt_rn((double)d), s2), s1))
-                       : 0.0f;
+            nx2[p] = __double2float_rn(t2);
+            F[p] = (t1 > 0.0) ? __double2float_rn(__ddiv_rn(__dmul_rn(sqrt_d, t2), t1)) : 0.0f;
             popx[p] = pc;
         }
     }

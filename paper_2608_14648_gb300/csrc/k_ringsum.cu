@@ -90,10 +90,13 @@ __device__ __forceinline__ int run_len(int64_t nval, int64_t q0) {
     return r <= 0 ? 0 : (r >= RS_ROWS ? RS_ROWS : (int)r);
 }
 
-// Shared-memory layout of one CTA (ns slots of sb bytes per consumer warp).
+// Shared-memory layout of one CTA: ns slots per consumer warp, each holding
+// up to R rows of rb bytes (small rows are batched so that one barrier round
+// trip covers about a kilobyte).
 struct RingLayout {
-    int ns, sb;
-    __host__ __device__ size_t ring_bytes() const { return (size_t)RS_CW * ns * sb; }
+    int ns, R, rb;
+    __host__ __device__ size_t slot_bytes() const { return (size_t)R * rb; }
+    __host__ __device__ size_t ring_bytes() const { return (size_t)RS_CW * ns * slot_bytes(); }
     __host__ __device__ size_t bytes() const {
         return ring_bytes() + (size_t)2 * RS_CW * ns * 8 + (size_t)RS_CW * RS_ROWS * 4 + 2 * RS_CW * 4;
     }
@@ -101,10 +104,10 @@ struct RingLayout {
 
 // Producer and teardown shared by every row type.  A consumer warp calls
 // cons.start(q0, cnt, lane) before the first row of its run (positions q0 ..
-// q0 + cnt - 1), cons.row(i, slot, lane) for its i-th row (in shared memory),
+// q0 + cnt - 1), cons.row(i, row, lane) for its i-th row (in shared memory),
 // and cons.finish(lane) after the last.
 template <typename Consumer>
-__device__ __forceinline__ void ring_run(const uint8_t *__restrict__ rows, uint32_t rb,
+__device__ __forceinline__ void ring_run(const uint8_t *__restrict__ rows,
                                          const int32_t *__restrict__ perm, int64_t nval,
                                          RingLayout L, volatile int32_t *flag, Consumer &cons) {
     extern __shared__ __align__(128) uint8_t rs_smem[];
@@ -112,10 +115,12 @@ __device__ __forceinline__ void ring_run(const uint8_t *__restrict__ rows, uint3
     uint64_t *full = reinterpret_cast<uint64_t *>(rs_smem + L.ring_bytes());
     uint64_t *empty = full + RS_CW * L.ns;
     int32_t *sperm = reinterpret_cast<int32_t *>(empty + RS_CW * L.ns);
-    int32_t *issued = sperm + RS_CW * RS_ROWS;
-    int32_t *consumed = issued + RS_CW;
+    int32_t *issued = sperm + RS_CW * RS_ROWS;  // slots filled, per stream
+    int32_t *consumed = issued + RS_CW;         // slots released, per stream
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int64_t qbase = (int64_t)blockIdx.x * RS_CW * RS_ROWS;
+    const uint32_t rb = (uint32_t)L.rb;
+    const size_t sb = L.slot_bytes();
 
     if (threadIdx.x == 0) {
         for (int i = 0; i < RS_CW * L.ns; ++i) {
@@ -138,48 +143,56 @@ __device__ __forceinline__ void ring_run(const uint8_t *__restrict__ rows, uint3
         __syncwarp();
         if (lane < RS_CW) {
             const int w = lane;
-            const int64_t q0 = qbase + (int64_t)w * RS_ROWS;
-            const int cnt = run_len(nval, q0);
-            int i = 0;
-            for (; i < cnt; ++i) {
-                const int s = i % L.ns;
-                const uint32_t ph = (uint32_t)(i / L.ns) & 1u;
+            const int cnt = run_len(nval, qbase + (int64_t)w * RS_ROWS);
+            int j = 0, s = 0;
+            uint32_t ph = 0;
+            for (int i0 = 0; i0 < cnt; i0 += L.R, ++j) {
+                const int nr = min(L.R, cnt - i0);
                 const uint32_t fb = su32(full + w * L.ns + s);
                 if (!bar_wait(su32(empty + w * L.ns + s), ph ^ 1u, flag)) break;
-                bar_arrive_tx(fb, rb);
-                bulk_g2s(su32(ring + ((size_t)w * L.ns + s) * L.sb),
-                         rows + (size_t)sperm[w * RS_ROWS + i] * rb, rb, fb);
+                bar_arrive_tx(fb, (uint32_t)nr * rb);
+                uint8_t *dst = ring + ((size_t)w * L.ns + s) * sb;
+                for (int r = 0; r < nr; ++r)
+                    bulk_g2s(su32(dst + (size_t)r * rb), rows + (size_t)sperm[w * RS_ROWS + i0 + r] * rb, rb, fb);
+                if (++s == L.ns) {
+                    s = 0;
+                    ph ^= 1u;
+                }
             }
-            issued[w] = i;
+            issued[w] = j;
         }
     } else {  // ------------------------------------------------------ consumers
         const int w = warp;
-        const int64_t q0 = qbase + (int64_t)w * RS_ROWS;
-        const int cnt = run_len(nval, q0);
-        int i = 0;
+        const int cnt = run_len(nval, qbase + (int64_t)w * RS_ROWS);
+        int j = 0;
         if (cnt > 0) {
-            cons.start(q0, cnt, lane);
-            for (; i < cnt; ++i) {
-                const int s = i % L.ns;
-                const uint32_t ph = (uint32_t)(i / L.ns) & 1u;
+            cons.start(qbase + (int64_t)w * RS_ROWS, cnt, lane);
+            int s = 0;
+            uint32_t ph = 0;
+            for (int i0 = 0; i0 < cnt; i0 += L.R, ++j) {
+                const int nr = min(L.R, cnt - i0);
                 const bool ok = bar_wait(su32(full + w * L.ns + s), ph, flag);
                 if (!__all_sync(0xffffffffu, ok)) break;
-                cons.row(i, ring + ((size_t)w * L.ns + s) * L.sb, lane);
+                const uint8_t *src = ring + ((size_t)w * L.ns + s) * sb;
+                for (int r = 0; r < nr; ++r) cons.row(i0 + r, src + (size_t)r * rb, lane);
                 __syncwarp();
                 if (lane == 0) bar_arrive(su32(empty + w * L.ns + s));
+                if (++s == L.ns) {
+                    s = 0;
+                    ph ^= 1u;
+                }
             }
             cons.finish(lane);
         }
-        if (lane == 0) consumed[w] = i;
+        if (lane == 0) consumed[w] = j;
     }
     __syncthreads();
-    // copies issued but never consumed (only after a wait gave up): let them land
+    // slots filled but never released (only after a wait gave up): let their
+    // copies land before the CTA's shared memory goes away
     if (warp == RS_CW && lane < RS_CW) {
         const int w = lane;
-        for (int i = consumed[w]; i < issued[w]; ++i) {
-            const int s = i % L.ns;
-            if (!bar_wait_drain(su32(full + w * L.ns + s), (uint32_t)(i / L.ns) & 1u)) break;
-        }
+        for (int j = consumed[w]; j < issued[w]; ++j)
+            if (!bar_wait_drain(su32(full + w * L.ns + j % L.ns), (uint32_t)(j / L.ns) & 1u)) break;
     }
 }
 
@@ -262,7 +275,7 @@ __global__ void __launch_bounds__(RS_THREADS) ring_sum_float_kernel(
     cons.S = S;
     cons.stride = stride;
     cons.d = d;
-    ring_run(static_cast<const uint8_t *>(X), (uint32_t)d * (BF16 ? 2u : 4u), perm, nval, L, flag, cons);
+    ring_run(static_cast<const uint8_t *>(X), perm, nval, L, flag, cons);
 }
 
 // ------------------------------------------------------------- 1-bit rows
@@ -319,15 +332,16 @@ struct Rbq1Cons {
             cur = c;
         }
         usum += fq;
+        const uint32_t lm = 1u << lane;
         const uint4 *w4 = reinterpret_cast<const uint4 *>(slot);
 #pragma unroll
         for (int g = 0; g < WM / 4; ++g) {
             if (4 * g < W) {
                 const uint4 wv = w4[g];  // broadcast: every lane reads the same 16 bytes
-                if ((wv.x >> lane) & 1u) acc[4 * g + 0] += fq;
-                if ((wv.y >> lane) & 1u) acc[4 * g + 1] += fq;
-                if ((wv.z >> lane) & 1u) acc[4 * g + 2] += fq;
-                if ((wv.w >> lane) & 1u) acc[4 * g + 3] += fq;
+                add_if_bit(acc[4 * g + 0], wv.x, lm, fq);
+                add_if_bit(acc[4 * g + 1], wv.y, lm, fq);
+                add_if_bit(acc[4 * g + 2], wv.z, lm, fq);
+                add_if_bit(acc[4 * g + 3], wv.w, lm, fq);
             }
         }
     }
@@ -348,13 +362,14 @@ __global__ void __launch_bounds__(RS_THREADS) ring_sum_rbq1_kernel(
     cons.T = T;
     cons.d = d;
     cons.W = (d + 31) >> 5;
-    ring_run(reinterpret_cast<const uint8_t *>(codes), (uint32_t)cons.W * 4u, perm, nval, L, flag, cons);
+    ring_run(reinterpret_cast<const uint8_t *>(codes), perm, nval, L, flag, cons);
 }
 
 bool ring_layout(uint32_t rb, RingLayout &L) {
     if (rb == 0 || rb % 16 != 0) return false;
-    L.sb = (int)rb;
-    L.ns = (int)std::min<size_t>(RS_MAX_SLOTS, RS_RING_BYTES / ((size_t)RS_CW * rb));
+    L.rb = (int)rb;
+    L.R = (int)std::max<uint32_t>(1u, std::min<uint32_t>(8u, 1024u / rb));
+    L.ns = (int)std::min<size_t>(RS_MAX_SLOTS, RS_RING_BYTES / ((size_t)RS_CW * L.slot_bytes()));
     return L.ns >= 2;
 }
 

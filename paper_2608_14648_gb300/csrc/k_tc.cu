@@ -64,12 +64,15 @@ constexpr int tc_threads() { return 64 + epi_threads<NH>(); }
 // one row's state for the merge: the screen list, or (best, index)
 template <int MODE>
 constexpr int merge_words() { return MODE == MODE_SCREEN ? 2 * TCAND + 2 : 2; }
-// 1024-byte alignment slack, the stages, barriers + TMEM slot (352 bytes), and
-// the merge buffer: slices 1..NH-1 publish, double-buffered by point tile
+// Per-centroid epilogue records of one centroid tile (256 columns): 4 KiB,
+// double-buffered by job.
+constexpr int REC_BYTES = 4096;
+// 1024-byte alignment slack, the stages, barriers + TMEM slot (352 bytes), the
+// merge buffer (slices 1..NH-1 publish) and the record buffers.
 template <int MODE, int NH>
 constexpr size_t tc_smem_bytes() {
     return 1024 + (size_t)STAGES * (A_STAGE + B_STAGE) + 512 +
-           (size_t)2 * (NH - 1) * BM * merge_words<MODE>() * 4;
+           (size_t)(NH - 1) * BM * merge_words<MODE>() * 4 + 2 * REC_BYTES;
 }
 
 struct TcParams {
@@ -406,10 +409,46 @@ __global__ void __launch_bounds__(tc_threads<NH>(), 1)
         const int q = warp & 3;          // TMEM lane quarter this warp may access
         const int slice = e >> 2;        // which SW of the 256 columns
         const int rin = q * 32 + lane;   // row within the point tile
-        uint32_t *merge = reinterpret_cast<uint32_t *>(tmem_slot + 64);  // [2][NH-1][BM][MW]
+        uint32_t *merge = reinterpret_cast<uint32_t *>(tmem_slot + 64);  // [NH-1][BM][MW]
+        // Records of the job's 256 centroids (SCREEN: 128 cinfo + 128 cinfoz
+        // pairs; RBQ1: 128 rinfo + 128 rinfoq pairs; SQ8: 256 nc), copied into
+        // shared memory at the start of each job from registers that were
+        // loaded one job ahead, so the per-column reads are shared-memory
+        // broadcasts.  Buffer (job & 1) is rewritten only after every epilogue
+        // thread has passed the next job's barrier, i.e. finished reading it.
+        uint8_t *rec_base = reinterpret_cast<uint8_t *>(merge + (NH - 1) * BM * MW);
+        const int te = threadIdx.x - 64;  // 0 .. epi_threads - 1
+        float4 pre4 = make_float4(0.f, 0.f, 0.f, 0.f);
+        float2 pre2 = make_float2(0.f, 0.f);
+        int32_t pre1 = 0;
+        auto rec_load = [&](int ctn) {
+            if (MODE == MODE_SCREEN) {
+                if (te < 128) pre4 = __ldg(p.cinfo + ctn * 128 + te);
+                else if (te < 256) pre2 = __ldg(p.cinfoz + ctn * 128 + (te - 128));
+            } else if (MODE == MODE_RBQ1) {
+                if (te < 128) pre4 = __ldg(p.rinfo + ctn * 128 + te);
+                else if (te < 256) pre4 = __ldg(p.rinfoq + ctn * 128 + (te - 128));
+            } else {
+                if (te < 256) pre1 = __ldg(p.nc + ctn * 256 + te);
+            }
+        };
+        auto rec_store = [&](uint32_t buf) {
+            uint8_t *rb = rec_base + buf * REC_BYTES;
+            if (MODE == MODE_SCREEN) {
+                if (te < 128) reinterpret_cast<float4 *>(rb)[te] = pre4;
+                else if (te < 256) reinterpret_cast<float2 *>(rb + 2048)[te - 128] = pre2;
+            } else if (MODE == MODE_RBQ1) {
+                if (te < 256) reinterpret_cast<float4 *>(rb)[te] = pre4;
+            } else {
+                if (te < 256) reinterpret_cast<int32_t *>(rb)[te] = pre1;
+            }
+        };
+        rec_load(0);
+        // A warp whose barrier wait gave up stops computing but keeps taking part
+        // in the named barriers, so the other epilogue warps never wait on it.
+        bool dead = false;
         uint32_t job = 0;
-        uint32_t tile = 0;
-        for (int64_t rt = blockIdx.x; rt < p.nrt; rt += gridDim.x, ++tile) {
+        for (int64_t rt = blockIdx.x; rt < p.nrt; rt += gridDim.x) {
             const int64_t row = rt * BM + rin;
             const bool valid = row < p.n;
             ScreenRow sr;
@@ -429,14 +468,21 @@ __global__ void __launch_bounds__(tc_threads<NH>(), 1)
             }
             for (int ct = 0; ct < p.nct; ++ct, ++job) {
                 const uint32_t b = job & 1u, bph = (job >> 1) & 1u;
-                const bool ok = mbar_wait(tfull_bar(b), bph, abort_flag);
-                if (!__all_sync(0xffffffffu, ok)) goto epi_done;
+                bool ok = true;
+                if (!dead) ok = mbar_wait(tfull_bar(b), bph, abort_flag);
+                dead = dead || !__all_sync(0xffffffffu, ok);
+                rec_store(b);
+                asm volatile("bar.sync 2, %0;" ::"n"(epi_threads<NH>()) : "memory");
+                rec_load(ct + 1 < p.nct ? ct + 1 : 0);
+                if (dead) continue;
                 tc_fence_after();
+                const uint8_t *rbuf = rec_base + b * REC_BYTES;
                 const uint32_t taddr = tmem + ((uint32_t)(q * 32) << 16) + b * BN + slice * SW;
                 const int jh = ct * BN + slice * SW;
 #pragma unroll 1
                 for (int c = 0; c < SW / 32; ++c) {
                     const int j0 = jh + c * 32;
+                    const int cc = slice * SW + c * 32;  // column offset within the tile
                     if (j0 >= p.k) break;  // warp-uniform
                     uint32_t v[32];
                     tmem_ld32(taddr + c * 32, v);
@@ -452,8 +498,8 @@ __global__ void __launch_bounds__(tc_threads<NH>(), 1)
                             cl[g] = INFINITY;
 #pragma unroll
                             for (int i = 8 * g; i < 8 * g + 8; i += 2) {
-                                const float4 ci = __ldg(p.cinfo + ((j0 + i) >> 1));
-                                const float2 cz = __ldg(p.cinfoz + ((j0 + i) >> 1));
+                                const float4 ci = reinterpret_cast<const float4 *>(rbuf)[(cc + i) >> 1];
+                                const float2 cz = reinterpret_cast<const float2 *>(rbuf + 2048)[(cc + i) >> 1];
                                 const float2 acc = make_float2(__uint_as_float(v[i]), __uint_as_float(v[i + 1]));
                                 const float2 m = ffma2(make_float2(-2.0f, -2.0f), acc, make_float2(ci.x, ci.y));
                                 const float2 w = ffma2(make_float2(a2, a2), make_float2(ci.z, ci.w), cz);
@@ -483,7 +529,7 @@ __global__ void __launch_bounds__(tc_threads<NH>(), 1)
 #pragma unroll
                         for (int i = 0; i < 32; ++i) {
                             const int32_t dot = __float2int_rn(__uint_as_float(v[i]));
-                            const int32_t dd = nxr + __ldg(p.nc + j0 + i) - 2 * dot;
+                            const int32_t dd = nxr + reinterpret_cast<const int32_t *>(rbuf)[cc + i] - 2 * dot;
                             if (dd < best) {
                                 best = dd;
                                 besti = j0 + i;
@@ -505,8 +551,8 @@ __global__ void __launch_bounds__(tc_threads<NH>(), 1)
                             gi[g] = 0x7fffffff;
 #pragma unroll
                             for (int i = 8 * g; i < 8 * g + 8; i += 2) {
-                                const float4 bs = __ldg(p.rinfo + ((j0 + i) >> 1));
-                                const float4 qn = __ldg(p.rinfoq + ((j0 + i) >> 1));
+                                const float4 bs = reinterpret_cast<const float4 *>(rbuf)[(cc + i) >> 1];
+                                const float4 qn = reinterpret_cast<const float4 *>(rbuf)[128 + ((cc + i) >> 1)];
                                 // packed pairs; every product here feeds an explicit fma
                                 // (no separate multiply-add the compiler could fuse)
                                 const float2 P2 = fsub2(
@@ -541,8 +587,11 @@ __global__ void __launch_bounds__(tc_threads<NH>(), 1)
                 mbar_arrive(tempty_bar(b));
             }
             // merge the column slices of each row: slices 1.. publish, slice 0 finishes
+            // (single buffer: a publisher rewrites its slot only at the end of
+            // the next point tile, after slice 0 has passed that tile's first
+            // job barrier, i.e. after it has read this one)
             if (slice > 0) {
-                uint32_t *slot = merge + (((tile & 1u) * (NH - 1) + (slice - 1)) * BM + rin) * MW;
+                uint32_t *slot = merge + ((slice - 1) * BM + rin) * MW;
                 if (MODE == MODE_SCREEN) {
 #pragma unroll
                     for (int t = 0; t < TCAND; ++t) {
@@ -560,11 +609,11 @@ __global__ void __launch_bounds__(tc_threads<NH>(), 1)
                 }
             }
             asm volatile("bar.sync 1, %0;" ::"n"(epi_threads<NH>()) : "memory");
-            if (slice == 0 && valid) {
+            if (slice == 0 && valid && !dead) {
                 // slices in increasing column order; ties resolve to the lower index
 #pragma unroll
                 for (int h = 1; h < NH; ++h) {
-                    const uint32_t *slot = merge + (((tile & 1u) * (NH - 1) + (h - 1)) * BM + rin) * MW;
+                    const uint32_t *slot = merge + ((h - 1) * BM + rin) * MW;
                     if (MODE == MODE_SCREEN) {
                         sr.umin = fminf(sr.umin, __uint_as_float(slot[2 * TCAND]));
                         sr.lev = fminf(sr.lev, __uint_as_float(slot[2 * TCAND + 1]));
@@ -613,7 +662,6 @@ __global__ void __launch_bounds__(tc_threads<NH>(), 1)
                 }
             }
         }
-    epi_done:;
     }
     tc_fence_before();
     __syncthreads();
@@ -627,37 +675,65 @@ __global__ void __launch_bounds__(tc_threads<NH>(), 1)
 
 // ------------------------------------------------------------- preparation
 // fp32 points -> bf16 screening copy (row stride dp) and per-row
-// (||x~||, ||x~ - x||), both rounded up.  One warp per row.
+// (||x~||, ||x~ - x||), both rounded up.  One warp per row.  The squares are
+// summed in fp32 (each lane sequentially, then an xor tree): a sum of m
+// non-negative terms carries a relative error below (m - 1) 2^-24 / (1 -
+// (m - 1) 2^-24), so the sums are scaled up by 1 + (m + 2) 2^-23 (rounded
+// up) before the upward-rounded square root.  x~_i - x_i is exact in fp32.
+__device__ __forceinline__ float sumsq_upper_norm(float s, int terms) {
+    const float grow = 1.0f + (float)(terms + 2) * 0x1p-23f;
+    return __fsqrt_ru(__fmul_ru(s, grow));
+}
+
+constexpr int PREP_UNROLL = 8;
+
 __global__ void screen_prep_f32_kernel(const float *__restrict__ X, int64_t n, int d, int dp,
                                        __nv_bfloat16 *__restrict__ xs, float2 *__restrict__ xinfo,
                                        unsigned int *__restrict__ rho_max_bits) {
     const int lane = threadIdx.x & 31;
     const int64_t warp = (blockIdx.x * (int64_t)blockDim.x + threadIdx.x) >> 5;
     const int64_t nw = ((int64_t)gridDim.x * blockDim.x) >> 5;
+    const int W = (d + 31) >> 5;
+    const int terms = W + 5;  // longest chain of roundings: per-lane terms + 5 tree levels
+    float rho_local = 0.0f;
     for (int64_t r = warp; r < n; r += nw) {
-        double a2 = 0.0, r2 = 0.0;
-        for (int i = lane; i < d; i += 32) {
-            const float x = X[r * d + i];
-            const __nv_bfloat16 xb = __float2bfloat16_rn(x);
-            xs[r * dp + i] = xb;
-            const double xf = (double)__bfloat162float(xb);
-            a2 += xf * xf;
-            r2 += (xf - (double)x) * (xf - (double)x);
+        float a2 = 0.0f, r2 = 0.0f;
+        for (int w0 = 0; w0 < W; w0 += PREP_UNROLL) {
+            float v[PREP_UNROLL];
+#pragma unroll
+            for (int u = 0; u < PREP_UNROLL; ++u) {
+                const int i = 32 * (w0 + u) + lane;
+                v[u] = (i < d) ? __ldg(X + r * d + i) : 0.0f;
+            }
+#pragma unroll
+            for (int u = 0; u < PREP_UNROLL; ++u) {
+                const int i = 32 * (w0 + u) + lane;
+                if (i < d) {
+                    const __nv_bfloat16 xb = __float2bfloat16_rn(v[u]);
+                    xs[r * dp + i] = xb;
+                    const float xf = __bfloat162float(xb);
+                    const float e = __fsub_rn(xf, v[u]);
+                    a2 = __fmaf_rn(xf, xf, a2);
+                    r2 = __fmaf_rn(e, e, r2);
+                }
+            }
         }
 #pragma unroll
         for (int o = 16; o > 0; o >>= 1) {
-            a2 += __shfl_xor_sync(0xffffffffu, a2, o);
-            r2 += __shfl_xor_sync(0xffffffffu, r2, o);
+            a2 = __fadd_rn(a2, __shfl_xor_sync(0xffffffffu, a2, o));
+            r2 = __fadd_rn(r2, __shfl_xor_sync(0xffffffffu, r2, o));
         }
         if (lane == 0) {
-            const float an = __double2float_ru(sqrt(a2) * (1.0 + 1e-6));
-            const float rn = __double2float_ru(sqrt(r2) * (1.0 + 1e-6));
+            const float an = sumsq_upper_norm(a2, terms);
+            const float rn = sumsq_upper_norm(r2, terms);
             xinfo[r] = make_float2(an, rn);
             // ratio ||x~ - x|| / ||x~|| (rounded up); x~ = 0 only when x = 0
             const float rho = an > 0.0f ? __fdiv_ru(rn, an) : 0.0f;
-            atomicMax(rho_max_bits, __float_as_uint(rho));  // non-negative: bits order as values
+            rho_local = (rho == rho) ? fmaxf(rho_local, rho) : INFINITY;  // NaN (inf data): no bound
         }
     }
+    // one atomic per warp; non-negative floats order like their bit patterns
+    if (lane == 0 && rho_local > 0.0f) atomicMax(rho_max_bits, __float_as_uint(rho_local));
 }
 
 // bf16 points: optional padded copy (when the row stride is not a multiple of
@@ -667,17 +743,18 @@ __global__ void screen_prep_bf16_kernel(const uint16_t *__restrict__ X, int64_t 
     const int lane = threadIdx.x & 31;
     const int64_t warp = (blockIdx.x * (int64_t)blockDim.x + threadIdx.x) >> 5;
     const int64_t nw = ((int64_t)gridDim.x * blockDim.x) >> 5;
+    const int terms = (d + 31) / 32 + 5;
     for (int64_t r = warp; r < n; r += nw) {
-        double a2 = 0.0;
+        float a2 = 0.0f;
         for (int i = lane; i < d; i += 32) {
             const uint16_t v = X[r * d + i];
             if (xs) xs[r * dp + i] = v;
-            const double xf = (double)__uint_as_float(((uint32_t)v) << 16);
-            a2 += xf * xf;
+            const float xf = __uint_as_float(((uint32_t)v) << 16);
+            a2 = __fmaf_rn(xf, xf, a2);
         }
 #pragma unroll
-        for (int o = 16; o > 0; o >>= 1) a2 += __shfl_xor_sync(0xffffffffu, a2, o);
-        if (lane == 0) xinfo[r] = make_float2(__double2float_ru(sqrt(a2) * (1.0 + 1e-6)), 0.0f);
+        for (int o = 16; o > 0; o >>= 1) a2 = __fadd_rn(a2, __shfl_xor_sync(0xffffffffu, a2, o));
+        if (lane == 0) xinfo[r] = make_float2(sumsq_upper_norm(a2, terms), 0.0f);
     }
 }
 

@@ -309,8 +309,6 @@ cudaError_t launch_rbq1_fq(const float *F, const int32_t *perm, const int64_t *o
     return launched();
 }
 
-constexpr int RB_WORDS = 32;  // code words per pass (1024 dimensions)
-
 // -------------------------------------------- chunked segmented sums (load balanced)
 // Warps take CH_ROWS consecutive members of the cluster-sorted order, so
 // every warp has the same work whatever the cluster sizes.  A warp adds its
@@ -381,27 +379,56 @@ __global__ void __launch_bounds__(CH_WARPS * 32) chunk_sum_float_kernel(
 }
 
 // 1-bit codes -> int64 accumulators T[k][d+1] (column d holds U = sum Fq);
-// fqs in the sorted order.
+// fqs in the sorted order.  Lane l holds dimension l of each code word.  A
+// warp's member ids, cluster ids and weights are read lane-parallel up
+// front; the member rows (W words, lane w loads word w) are read RB_DEPTH
+// rows ahead into a register ring, and each row's words reach every lane by
+// shuffles, so the loads of later rows overlap the sums of earlier ones.
+constexpr int RB_DEPTH = 8;
+
+__device__ __forceinline__ int pick4(const int (&a)[4], int i) {
+    const int t = i >> 5;
+    const int v = t == 0 ? a[0] : t == 1 ? a[1] : t == 2 ? a[2] : a[3];
+    return __shfl_sync(0xffffffffu, v, i & 31);
+}
+__device__ __forceinline__ int64_t pick4(const int64_t (&a)[4], int i) {
+    const int t = i >> 5;
+    const int64_t v = t == 0 ? a[0] : t == 1 ? a[1] : t == 2 ? a[2] : a[3];
+    return __shfl_sync(0xffffffffu, v, i & 31);
+}
+
+template <int WM>
 __global__ void __launch_bounds__(CH_WARPS * 32) chunk_sum_rbq1_kernel(
     const uint32_t *__restrict__ codes, const int64_t *__restrict__ fqs, int d,
     const int32_t *__restrict__ perm, const int32_t *__restrict__ scl,
     const int64_t *__restrict__ offsets, int k, unsigned long long *__restrict__ T) {
+    static_assert(CH_ROWS == 128, "pick4 covers 4 x 32 positions");
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int64_t nval = offsets[k];
     const int64_t q0 = ((int64_t)blockIdx.x * CH_WARPS + warp) * CH_ROWS;
     if (q0 >= nval) return;
-    const int64_t q1 = min(nval, q0 + CH_ROWS);
+    const int cnt = (int)(nval - q0 < CH_ROWS ? nval - q0 : CH_ROWS);
     const int W = (d + 31) >> 5;
-    for (int w0 = 0; w0 < W; w0 += RB_WORDS) {
-        const int nw = min(RB_WORDS, W - w0);
-        int64_t acc[RB_WORDS];
+    const uint32_t lm = 1u << lane;
+    int pp[4], cc[4];
+    int64_t ff[4];
 #pragma unroll
-        for (int t = 0; t < RB_WORDS; ++t) acc[t] = 0;
+    for (int t = 0; t < 4; ++t) {
+        const int i = lane + 32 * t;
+        pp[t] = i < cnt ? perm[q0 + i] : 0;
+        cc[t] = i < cnt ? scl[q0 + i] : -1;
+        ff[t] = i < cnt ? fqs[q0 + i] : 0;
+    }
+    for (int w0 = 0; w0 < W; w0 += WM) {
+        const int nw = min(WM, W - w0);
+        int64_t acc[WM];
+#pragma unroll
+        for (int t = 0; t < WM; ++t) acc[t] = 0;
         int64_t usum = 0;
-        int cur = scl[q0];
+        int cur = pick4(cc, 0);
         auto flush = [&](int c) {
 #pragma unroll
-            for (int t = 0; t < RB_WORDS; ++t) {
+            for (int t = 0; t < WM; ++t) {
                 const int col = 32 * (w0 + t) + lane;
                 if (t < nw && col < d && acc[t])
                     atomicAdd(T + (int64_t)c * (d + 1) + col, (unsigned long long)acc[t]);
@@ -410,20 +437,35 @@ __global__ void __launch_bounds__(CH_WARPS * 32) chunk_sum_rbq1_kernel(
             if (w0 == 0 && lane == 0 && usum) atomicAdd(T + (int64_t)c * (d + 1) + d, (unsigned long long)usum);
             usum = 0;
         };
-        for (int64_t q = q0; q < q1; ++q) {
-            const int c = scl[q];
-            const int64_t p = perm[q];
-            const int64_t fq = __ldg(fqs + q);
-            const uint32_t mine = (lane < nw) ? __ldg(codes + p * W + w0 + lane) : 0u;
-            if (c != cur) {
-                flush(cur);
-                cur = c;
-            }
-            usum += fq;
+        uint32_t buf[RB_DEPTH];
 #pragma unroll
-            for (int t = 0; t < RB_WORDS; ++t) {
-                const uint32_t word = __shfl_sync(0xffffffffu, mine, t);
-                if ((word >> lane) & 1u) acc[t] += fq;
+        for (int r = 0; r < RB_DEPTH; ++r) {
+            const int p = pick4(pp, r);
+            buf[r] = (r < cnt && lane < nw) ? __ldg(codes + (int64_t)p * W + w0 + lane) : 0u;
+        }
+        for (int i0 = 0; i0 < cnt; i0 += RB_DEPTH) {
+#pragma unroll
+            for (int r = 0; r < RB_DEPTH; ++r) {
+                const int i = i0 + r;
+                const uint32_t mine = buf[r];
+                const int in = i + RB_DEPTH;
+                const int pn = pick4(pp, in < CH_ROWS ? in : 0);
+                buf[r] = (in < cnt && lane < nw) ? __ldg(codes + (int64_t)pn * W + w0 + lane) : 0u;
+                if (i < cnt) {  // warp-uniform
+                    const int c = pick4(cc, i);
+                    const int64_t fq = pick4(ff, i);
+                    if (c != cur) {
+                        flush(cur);
+                        cur = c;
+                    }
+                    usum += fq;
+#pragma unroll
+                    for (int t = 0; t < WM; ++t) {
+                        if (t < nw) {
+                            add_if_bit(acc[t], __shfl_sync(0xffffffffu, mine, t), lm, fq);
+                        }
+                    }
+                }
             }
         }
         flush(cur);
@@ -460,8 +502,17 @@ cudaError_t launch_chunk_sum_rbq1(const uint32_t *codes, const int64_t *fq, int6
                                   const int32_t *perm, const int32_t *scl, const int64_t *offsets,
                                   int k, int64_t *T, cudaStream_t st) {
     if (n == 0) return cudaSuccess;
-    chunk_sum_rbq1_kernel<<<chunk_blocks(n), CH_WARPS * 32, 0, st>>>(
-        codes, fq, d, perm, scl, offsets, k, reinterpret_cast<unsigned long long *>(T));
+    const int W = (d + 31) >> 5;
+    auto T64 = reinterpret_cast<unsigned long long *>(T);
+    const unsigned g = chunk_blocks(n);
+    if (W <= 8)
+        chunk_sum_rbq1_kernel<8><<<g, CH_WARPS * 32, 0, st>>>(codes, fq, d, perm, scl, offsets, k, T64);
+    else if (W <= 16)
+        chunk_sum_rbq1_kernel<16><<<g, CH_WARPS * 32, 0, st>>>(codes, fq, d, perm, scl, offsets, k, T64);
+    else if (W <= 24)
+        chunk_sum_rbq1_kernel<24><<<g, CH_WARPS * 32, 0, st>>>(codes, fq, d, perm, scl, offsets, k, T64);
+    else
+        chunk_sum_rbq1_kernel<32><<<g, CH_WARPS * 32, 0, st>>>(codes, fq, d, perm, scl, offsets, k, T64);
     return launched();
 }
 

@@ -55,6 +55,17 @@ struct Carver {
 inline int words_of(int d) { return (d + 31) / 32; }
 inline int64_t cdiv(int64_t a, int64_t b) { return (a + b - 1) / b; }
 
+// acc += fq when (word & mask) != 0, as a predicated add (no branch); used
+// by the 1-bit decode-average sums.
+__device__ __forceinline__ void add_if_bit(int64_t &acc, uint32_t word, uint32_t mask, int64_t fq) {
+    asm("{\n\t.reg .pred p;\n\t"
+        "and.b32 %1, %1, %2;\n\t"
+        "setp.ne.u32 p, %1, 0;\n\t"
+        "@p add.s64 %0, %0, %3;\n\t}"
+        : "+l"(acc), "+r"(word)
+        : "r"(mask), "l"(fq));
+}
+
 // Per-centroid terms of the RBQ1 estimator (Eq. final:rabitq), one record
 // per centroid: SQ4 bias and scale multiplied by fl(1/sqrt(d)) (bd = b isd,
 // sd = s isd), the sum of codes, ||c - m||^2.

@@ -98,6 +98,52 @@ def test_update_f32_vs_oracle(skm):
     np.testing.assert_array_equal(C.cpu().numpy()[k - 1], C0.numpy()[k - 1])  # empty cluster kept
 
 
+def _skewed_assign(n, k, seed):
+    """60% of the points in cluster 0, the rest spread over 1..k-2 (k-1 stays
+    empty), and every 997th point outside [0, k) (skipped by the update)."""
+    g = torch.Generator().manual_seed(seed)
+    a = torch.randint(1, k - 1, (n,), generator=g, dtype=torch.int32)
+    a[torch.rand(n, generator=g) < 0.6] = 0
+    a[::997] = -1
+    return a
+
+
+@pytest.mark.parametrize("repr_name,n,d,k", [("f32", 70001, 128, 500), ("f32", 9000, 1536, 40),
+                                             ("bf16", 20011, 1024, 300), ("rbq1", 70001, 128, 500),
+                                             ("rbq1", 20011, 1024, 300)])
+def test_update_skewed_clusters(skm, repr_name, n, d, k):
+    """Runs of the sorted order that cross many small clusters and one giant
+    cluster shared by hundreds of runs; ragged last run; skipped points."""
+    X = _points(n, d, seed=n + d)
+    a = _skewed_assign(n, k, seed=d)
+    ok = (a >= 0).numpy()
+    C0 = X[:k].clone()
+    if repr_name == "rbq1":
+        r = skm.skm_quantize(skm.REPR_RBQ1, X.to(DEV))
+        pts = skm.rbq1_points(r, d)
+        h = _rbq1_host(r)
+        Cn, counts = skm.skm_update(pts, a.to(DEV), C0.to(DEV).clone())
+        Co, co = oracle.rbq1_update(h["codes"][ok], h["F"][ok], d, h["m"], pts.rbq1_exp,
+                                    a.numpy()[ok], C0.numpy())
+        np.testing.assert_array_equal(counts.cpu().numpy(), co)
+        np.testing.assert_array_equal(Cn.cpu().numpy(), Co)
+        return
+    if repr_name == "bf16":
+        Xb = X.to(torch.bfloat16)
+        pts = skm.Points(skm.REPR_BF16, Xb.view(torch.int16).to(DEV), d)
+        Co, co = oracle.update_bf16(Xb.view(torch.int16).numpy().view(np.uint16)[ok], a.numpy()[ok],
+                                    C0.numpy())
+    else:
+        pts = skm.Points(skm.REPR_F32, X.to(DEV), d)
+        Co, co = oracle.update_f32(X.numpy()[ok], a.numpy()[ok], C0.numpy())
+    Cn, counts = skm.skm_update(pts, a.to(DEV), C0.to(DEV).clone())
+    np.testing.assert_array_equal(counts.cpu().numpy(), co)
+    Cg = Cn.cpu().numpy().astype(np.float64)
+    rel = np.linalg.norm(Cg - Co, axis=1) / np.maximum(np.linalg.norm(Co, axis=1), 1e-30)
+    assert rel.max() <= 1e-4
+    np.testing.assert_array_equal(Cn.cpu().numpy()[k - 1], C0.numpy()[k - 1])  # empty cluster kept
+
+
 def test_fit_f32_tiny_workload(skm):
     spec = synth.WORKLOADS["tiny_f32"]
     X = synth.workload_points(spec, seed=0)
