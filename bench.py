@@ -33,6 +33,8 @@ N_POINTS, DIM, K, N_COMP = 1_000_000, 768, 1000, 2000
 METRIC = "k-means point·centroid distances/s per Lloyd iter (1 GB300); % of roofline"
 WORKLOAD = "emb1m_d768: N=1,000,000 x d=768 unit-norm GMM embeddings, k=1,000; fp32 + RabitQ 1-bit"
 SM_COUNT = 152
+# row ranges of the end-to-end step's host-to-device copy (overlapped with work)
+E2E_CHUNKS = 16
 # POPC results per clock per SM used for the 1-bit kernel's ALU roofline
 # (measured 15.9 on GB300 with a throughput probe).
 POPC_PER_CLK_SM = 16
@@ -301,9 +303,32 @@ def run_ours(args):
         Xd2 = torch.empty_like(X)
         Cd32 = torch.empty_like(C32)
         CdR = torch.empty_like(Cr)
-        pts2 = skm.Points(skm.REPR_F32, Xd2, DIM)  # screening copies rebuilt inside every call
-        wsA2 = skm.workspace(skm.OP_ASSIGN, pts2, K)
-        wsAR2 = skm.workspace(skm.OP_ASSIGN, skm.rbq1_points(q, DIM, e), K)
+        # The H2D copy of the points is cut into E2E_CHUNKS row ranges on a copy
+        # stream; each range is assigned (fp32: screening copy built inside the
+        # call; 1-bit: encoded, then assigned) and its fp32 cluster sums are
+        # added into fp64 partial sums (the sharded update form) as soon as it
+        # has landed, so the copy of later ranges overlaps the work on earlier
+        # ones.  The fp32 update is finalised after the last range; the 1-bit
+        # update needs the fixed-point exponent of every F and runs after it.
+        nchunk = E2E_CHUNKS
+        bounds = [(i * N_POINTS // nchunk, (i + 1) * N_POINTS // nchunk) for i in range(nchunk)]
+        cmax = max(b1 - b0 for b0, b1 in bounds)
+        W = (DIM + 31) // 32
+        codesE = torch.empty(N_POINTS, W, device=dev, dtype=torch.int32)
+        nx2E = torch.empty(N_POINTS, device=dev, dtype=torch.float32)
+        FE = torch.empty(N_POINTS, device=dev, dtype=torch.float32)
+        popxE = torch.empty(N_POINTS, device=dev, dtype=torch.int32)
+        mE = q["m"]
+        probe32 = skm.Points(skm.REPR_F32, Xd2[:cmax], DIM)
+        wsA2 = skm.workspace(skm.OP_ASSIGN, probe32, K)
+        wsAR2 = skm.workspace(skm.OP_ASSIGN, skm.Points(skm.REPR_RBQ1, codesE[:cmax], DIM, nx2E[:cmax],
+                                                        FE[:cmax], popxE[:cmax], mE, e), K)
+        wsQ2 = skm.workspace(skm.OP_QUANTIZE, probe32, 1)
+        part32e = torch.zeros(K, DIM, device=dev, dtype=torch.float64)
+        cnt32e = torch.zeros(K, device=dev, dtype=torch.int64)
+        wsU2 = skm.workspace(skm.OP_UPDATE, probe32, K)
+        copy_stream = torch.cuda.Stream()
+        landed = [torch.cuda.Event() for _ in range(nchunk)]
         h2d = X_host.numel() * 4 + 2 * K * DIM * 4
         d2h = 2 * N_POINTS * 4 + 2 * K * DIM * 4
         e2e_steps = max(2, min(args.steps, 5))
@@ -313,14 +338,29 @@ def run_ours(args):
         s0, s1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
         s0.record(stream)
         for _ in range(e2e_steps):
-            Xd2.copy_(X_host, non_blocking=True)
+            copy_stream.wait_stream(stream)  # the previous step is done with Xd2
+            with torch.cuda.stream(copy_stream):
+                for (b0, b1), ev in zip(bounds, landed):
+                    Xd2[b0:b1].copy_(X_host[b0:b1], non_blocking=True)
+                    ev.record(copy_stream)
             Cd32.copy_(C_host32, non_blocking=True)
             CdR.copy_(C_hostR, non_blocking=True)
-            qq = skm.skm_quantize(skm.REPR_RBQ1, Xd2, fit=False, m=q["m"])
-            pR2 = skm.rbq1_points(qq, DIM, e)
-            skm.skm_assign(pts2, Cd32, K, want_dist=False, ws=wsA2, out=a32)
-            skm.skm_update(pts2, a32, Cd32, counts=cnt32, ws=wsU32)
-            skm.skm_assign(pR2, CdR, K, want_dist=False, ws=wsAR2, out=aR)
+            part32e.zero_()
+            cnt32e.zero_()
+            for (b0, b1), ev in zip(bounds, landed):
+                stream.wait_event(ev)
+                Xc = Xd2[b0:b1]
+                pc = skm.Points(skm.REPR_F32, Xc, DIM)
+                skm.skm_assign(pc, Cd32, K, want_dist=False, ws=wsA2, out=a32[b0:b1])
+                skm.skm_update(pc, a32[b0:b1], None, counts=cnt32e, partial=part32e, ws=wsU2)
+                qc = skm.skm_quantize(skm.REPR_RBQ1, Xc, fit=False, m=mE, ws=wsQ2,
+                                      out={"codes": codesE[b0:b1], "nx2": nx2E[b0:b1], "F": FE[b0:b1],
+                                           "popx": popxE[b0:b1]})
+                skm.skm_assign(skm.rbq1_points(qc, DIM, e), CdR, K, want_dist=False, ws=wsAR2,
+                               out=aR[b0:b1])
+            skm.skm_update_finalize(skm.Points(skm.REPR_F32, Xd2, DIM), part32e, cnt32e, Cd32)
+            eE = skm.skm_rbq1_exponent(FE)
+            pR2 = skm.Points(skm.REPR_RBQ1, codesE, DIM, nx2E, FE, popxE, mE, eE)
             skm.skm_update(pR2, aR, CdR, counts=cntR, ws=wsUR)
             a_host[0].copy_(a32, non_blocking=True)
             a_host[1].copy_(aR, non_blocking=True)
@@ -336,8 +376,9 @@ def run_ours(args):
         e2e = {"value": world * 2.0 * N_POINTS * K * e2e_steps / (ems / 1e3), "unit": "distances/s",
                "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "steps": e2e_steps,
                "ms_per_step": ems / e2e_steps,
-               "path": "pinned host fp32 points -> H2D -> skm_quantize(RBQ1) -> skm_assign/skm_update "
-                       "(fp32, 1-bit) -> D2H assignments + centroids"}
+               "path": f"pinned host fp32 points -> H2D in {nchunk} row ranges on a copy stream, each "
+                       "range assigned (fp32) and encoded + assigned (1-bit) once it has landed -> "
+                       "skm_update (fp32, 1-bit) -> D2H assignments + centroids"}
 
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:

@@ -213,16 +213,20 @@ def skm_pca_fit(X, d_out, stream=None):
     return mean, P, w
 
 
-def skm_quantize(repr_, X, fit=True, b=None, s=None, m=None, stream=None):
-    """SQ8 -> dict(codes, b, s); RBQ1 -> dict(codes, m, nx2, F, popx)."""
+def skm_quantize(repr_, X, fit=True, b=None, s=None, m=None, stream=None, out=None, ws=None):
+    """SQ8 -> dict(codes, b, s); RBQ1 -> dict(codes, m, nx2, F, popx).
+    `out` may supply preallocated (contiguous) output tensors by those names."""
     n, d = X.shape
     dev = X.device
-    dummy = Points(REPR_F32, X, d)
-    ws = _ws(skm_workspace_size(OP_QUANTIZE, dummy, 1), dev)
+    out = out or {}
+    if ws is None:
+        dummy = Points(REPR_F32, X, d)
+        ws = _ws(skm_workspace_size(OP_QUANTIZE, dummy, 1), dev)
     if repr_ == REPR_SQ8:
         b = b if b is not None else torch.empty(d, device=dev, dtype=torch.float32)
         s = s if s is not None else torch.empty(d, device=dev, dtype=torch.float32)
-        codes = torch.empty(n, d, device=dev, dtype=torch.uint8)
+        codes = out.get("codes")
+        codes = codes if codes is not None else torch.empty(n, d, device=dev, dtype=torch.uint8)
         qp = QuantParams(int(fit), 0, b.data_ptr(), s.data_ptr(), None, None, None, None)
         _check(lib().skm_quantize(repr_, _ptr(X), n, d, ctypes.byref(qp), _ptr(codes), _ptr(ws), ws.numel(),
                                   _stream(stream)))
@@ -230,10 +234,17 @@ def skm_quantize(repr_, X, fit=True, b=None, s=None, m=None, stream=None):
     if repr_ == REPR_RBQ1:
         W = (d + 31) // 32
         m = m if m is not None else torch.empty(d, device=dev, dtype=torch.float32)
-        codes = torch.empty(n, W, device=dev, dtype=torch.int32)
-        nx2 = torch.empty(n, device=dev, dtype=torch.float32)
-        F = torch.empty(n, device=dev, dtype=torch.float32)
-        popx = torch.empty(n, device=dev, dtype=torch.int32)
+        def _o(name, shape, dt):
+            t = out.get(name)
+            if t is None:
+                return torch.empty(*shape, device=dev, dtype=dt)
+            if not t.is_contiguous() or tuple(t.shape) != tuple(shape) or t.dtype != dt:
+                raise ValueError(f"out[{name!r}] must be a contiguous {dt} tensor of shape {shape}")
+            return t
+        codes = _o("codes", (n, W), torch.int32)
+        nx2 = _o("nx2", (n,), torch.float32)
+        F = _o("F", (n,), torch.float32)
+        popx = _o("popx", (n,), torch.int32)
         qp = QuantParams(int(fit), 0, None, None, m.data_ptr(), nx2.data_ptr(), F.data_ptr(), popx.data_ptr())
         _check(lib().skm_quantize(repr_, _ptr(X), n, d, ctypes.byref(qp), _ptr(codes), _ptr(ws), ws.numel(),
                                   _stream(stream)))

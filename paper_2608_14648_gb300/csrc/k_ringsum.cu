@@ -280,14 +280,17 @@ __global__ void __launch_bounds__(RS_THREADS) ring_sum_float_kernel(
 
 // ------------------------------------------------------------- 1-bit rows
 // T[c][i] += Fq for every member with bit i set; T[c][d] += Fq (= U).
-// Lane l holds dimension l of every code word (t < WM words).
-template <int WM>
+// Lane l holds dimension l of each of the W = 4 W4 code words.  Inside a run
+// (at most RS_ROWS rows between flushes) Fq = hi 2^20 + lo is accumulated as
+// two 32-bit sums, which cannot overflow (Fq <= 2^37: sum lo < 2^27, sum hi
+// <= 2^24), so each (row, dimension) costs one test and two predicated adds.
+template <int W4>
 struct Rbq1Cons {
     const int32_t *scl;
     const int64_t *fqs;  // Fq in sorted order
     unsigned long long *T;
-    int d, W;
-    int64_t acc[WM];
+    int d;
+    uint32_t alo[4 * W4], ahi[4 * W4];
     int64_t usum;
     int cur;
     int64_t q0;
@@ -296,11 +299,12 @@ struct Rbq1Cons {
     int cnt;
     __device__ __forceinline__ void flush(int c, int lane) {
 #pragma unroll
-        for (int t = 0; t < WM; ++t) {
+        for (int t = 0; t < 4 * W4; ++t) {
             const int col = 32 * t + lane;
-            if (t < W && col < d && acc[t])
-                atomicAdd(T + (int64_t)c * (d + 1) + col, (unsigned long long)acc[t]);
-            acc[t] = 0;
+            const unsigned long long v = ((unsigned long long)ahi[t] << 20) + alo[t];
+            if (col < d && v) atomicAdd(T + (int64_t)c * (d + 1) + col, v);
+            alo[t] = 0;
+            ahi[t] = 0;
         }
         if (lane == 0 && usum) atomicAdd(T + (int64_t)c * (d + 1) + d, (unsigned long long)usum);
         usum = 0;
@@ -309,7 +313,10 @@ struct Rbq1Cons {
         q0 = q0_;
         cnt = cnt_;
 #pragma unroll
-        for (int t = 0; t < WM; ++t) acc[t] = 0;
+        for (int t = 0; t < 4 * W4; ++t) {
+            alo[t] = 0;
+            ahi[t] = 0;
+        }
         usum = 0;
         clw = lane < cnt ? __ldg(scl + q0 + lane) : -1;
         cln = 32 + lane < cnt ? __ldg(scl + q0 + 32 + lane) : -1;
@@ -332,23 +339,22 @@ struct Rbq1Cons {
             cur = c;
         }
         usum += fq;
+        const uint32_t flo = (uint32_t)fq & 0xfffffu, fhi = (uint32_t)(fq >> 20);
         const uint32_t lm = 1u << lane;
         const uint4 *w4 = reinterpret_cast<const uint4 *>(slot);
 #pragma unroll
-        for (int g = 0; g < WM / 4; ++g) {
-            if (4 * g < W) {
-                const uint4 wv = w4[g];  // broadcast: every lane reads the same 16 bytes
-                add_if_bit(acc[4 * g + 0], wv.x, lm, fq);
-                add_if_bit(acc[4 * g + 1], wv.y, lm, fq);
-                add_if_bit(acc[4 * g + 2], wv.z, lm, fq);
-                add_if_bit(acc[4 * g + 3], wv.w, lm, fq);
-            }
+        for (int g = 0; g < W4; ++g) {
+            const uint4 wv = w4[g];  // broadcast: every lane reads the same 16 bytes
+            add_if_bit2(alo[4 * g + 0], ahi[4 * g + 0], wv.x, lm, flo, fhi);
+            add_if_bit2(alo[4 * g + 1], ahi[4 * g + 1], wv.y, lm, flo, fhi);
+            add_if_bit2(alo[4 * g + 2], ahi[4 * g + 2], wv.z, lm, flo, fhi);
+            add_if_bit2(alo[4 * g + 3], ahi[4 * g + 3], wv.w, lm, flo, fhi);
         }
     }
     __device__ __forceinline__ void finish(int lane) { flush(cur, lane); }
 };
 
-template <int WM>
+template <int W4>
 __global__ void __launch_bounds__(RS_THREADS) ring_sum_rbq1_kernel(
     const uint32_t *__restrict__ codes, const int64_t *__restrict__ fqs, int d,
     const int32_t *__restrict__ perm, const int32_t *__restrict__ scl,
@@ -356,12 +362,11 @@ __global__ void __launch_bounds__(RS_THREADS) ring_sum_rbq1_kernel(
     int32_t *flag) {
     const int64_t nval = offsets[k];
     if ((int64_t)blockIdx.x * RS_CW * RS_ROWS >= nval) return;
-    Rbq1Cons<WM> cons;
+    Rbq1Cons<W4> cons;
     cons.scl = scl;
     cons.fqs = fqs;
     cons.T = T;
     cons.d = d;
-    cons.W = (d + 31) >> 5;
     ring_run(reinterpret_cast<const uint8_t *>(codes), perm, nval, L, flag, cons);
 }
 
@@ -446,18 +451,26 @@ cudaError_t launch_ring_sum_rbq1(const uint32_t *codes, const int64_t *fqs, int6
     const size_t smem = L.bytes();
     const unsigned g = ring_blocks(n);
     auto T64 = reinterpret_cast<unsigned long long *>(T);
-#define RS_CASE(WMV)                                                                                \
-    if (W <= WMV) {                                                                                 \
-        auto kern = ring_sum_rbq1_kernel<WMV>;                                                      \
+#define RS_CASE(W4V)                                                                                \
+    case W4V: {                                                                                     \
+        auto kern = ring_sum_rbq1_kernel<W4V>;                                                      \
         cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem); \
         if (e != cudaSuccess) return e;                                                             \
         kern<<<g, RS_THREADS, smem, st>>>(codes, fqs, d, perm, scl, offsets, k, T64, L, flag);       \
         return launched();                                                                          \
     }
-    RS_CASE(8)
-    RS_CASE(16)
-    RS_CASE(24)
-    RS_CASE(32)
+    switch (W / 4) {
+        RS_CASE(1)
+        RS_CASE(2)
+        RS_CASE(3)
+        RS_CASE(4)
+        RS_CASE(5)
+        RS_CASE(6)
+        RS_CASE(7)
+        RS_CASE(8)
+    default:
+        break;
+    }
 #undef RS_CASE
     return cudaErrorInvalidValue;
 }

@@ -421,18 +421,20 @@ __global__ void __launch_bounds__(CH_WARPS * 32) chunk_sum_rbq1_kernel(
     }
     for (int w0 = 0; w0 < W; w0 += WM) {
         const int nw = min(WM, W - w0);
-        int64_t acc[WM];
+        // Fq = hi 2^20 + lo as two 32-bit sums (at most CH_ROWS rows between
+        // flushes: sum lo < 2^27, sum hi <= 2^24)
+        uint32_t alo[WM], ahi[WM];
 #pragma unroll
-        for (int t = 0; t < WM; ++t) acc[t] = 0;
+        for (int t = 0; t < WM; ++t) alo[t] = ahi[t] = 0u;
         int64_t usum = 0;
         int cur = pick4(cc, 0);
         auto flush = [&](int c) {
 #pragma unroll
             for (int t = 0; t < WM; ++t) {
                 const int col = 32 * (w0 + t) + lane;
-                if (t < nw && col < d && acc[t])
-                    atomicAdd(T + (int64_t)c * (d + 1) + col, (unsigned long long)acc[t]);
-                acc[t] = 0;
+                const unsigned long long v = ((unsigned long long)ahi[t] << 20) + alo[t];
+                if (t < nw && col < d && v) atomicAdd(T + (int64_t)c * (d + 1) + col, v);
+                alo[t] = ahi[t] = 0u;
             }
             if (w0 == 0 && lane == 0 && usum) atomicAdd(T + (int64_t)c * (d + 1) + d, (unsigned long long)usum);
             usum = 0;
@@ -459,10 +461,11 @@ __global__ void __launch_bounds__(CH_WARPS * 32) chunk_sum_rbq1_kernel(
                         cur = c;
                     }
                     usum += fq;
+                    const uint32_t flo = (uint32_t)fq & 0xfffffu, fhi = (uint32_t)(fq >> 20);
 #pragma unroll
                     for (int t = 0; t < WM; ++t) {
                         if (t < nw) {
-                            add_if_bit(acc[t], __shfl_sync(0xffffffffu, mine, t), lm, fq);
+                            add_if_bit2(alo[t], ahi[t], __shfl_sync(0xffffffffu, mine, t), lm, flo, fhi);
                         }
                     }
                 }

@@ -55,15 +55,18 @@ struct Carver {
 inline int words_of(int d) { return (d + 31) / 32; }
 inline int64_t cdiv(int64_t a, int64_t b) { return (a + b - 1) / b; }
 
-// acc += fq when (word & mask) != 0, as a predicated add (no branch); used
-// by the 1-bit decode-average sums.
-__device__ __forceinline__ void add_if_bit(int64_t &acc, uint32_t word, uint32_t mask, int64_t fq) {
+// (lo, hi) += (flo, fhi) when (word & mask) != 0, as two predicated 32-bit
+// adds (no branch, no carry); used by the 1-bit decode-average sums, which
+// split each fixed-point weight as hi 2^20 + lo.
+__device__ __forceinline__ void add_if_bit2(uint32_t &lo, uint32_t &hi, uint32_t word, uint32_t mask,
+                                            uint32_t flo, uint32_t fhi) {
     asm("{\n\t.reg .pred p;\n\t"
-        "and.b32 %1, %1, %2;\n\t"
-        "setp.ne.u32 p, %1, 0;\n\t"
-        "@p add.s64 %0, %0, %3;\n\t}"
-        : "+l"(acc), "+r"(word)
-        : "r"(mask), "l"(fq));
+        "and.b32 %2, %2, %3;\n\t"
+        "setp.ne.u32 p, %2, 0;\n\t"
+        "@p add.u32 %0, %0, %4;\n\t"
+        "@p add.u32 %1, %1, %5;\n\t}"
+        : "+r"(lo), "+r"(hi), "+r"(word)
+        : "r"(mask), "r"(flo), "r"(fhi));
 }
 
 // Per-centroid terms of the RBQ1 estimator (Eq. final:rabitq), one record
