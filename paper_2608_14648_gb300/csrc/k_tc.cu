@@ -82,6 +82,7 @@ struct TcParams {
     int nct;  // centroid tiles
     int nkc;  // 64-wide k-slices
     const float4 *cinfo;  // SCREEN: per column pair (||c||^2 x2, h' x2), padded to 256
+    const float *hz;      // SCREEN: (max h', max z) over the centroids
     const float2 *cinfoz; // SCREEN: per column pair (z x2)
     const float2 *xinfo;  // SCREEN: per point (||x~||, ||x~ - x||)
     int32_t *cand;        // SCREEN: [n][TCAND + 1]
@@ -410,8 +411,8 @@ __global__ void __launch_bounds__(tc_threads<NH>(), 1)
         const int slice = e >> 2;        // which SW of the 256 columns
         const int rin = q * 32 + lane;   // row within the point tile
         uint32_t *merge = reinterpret_cast<uint32_t *>(tmem_slot + 64);  // [NH-1][BM][MW]
-        // Records of the job's 256 centroids (SCREEN: 128 cinfo + 128 cinfoz
-        // pairs; RBQ1: 128 rinfo + 128 rinfoq pairs; SQ8: 256 nc), copied into
+        // Records of the job's 256 centroids (SCREEN: 128 ||c||^2 pairs; RBQ1:
+        // 128 rinfo + 128 rinfoq pairs; SQ8: 256 nc), copied into
         // shared memory at the start of each job from registers that were
         // loaded one job ahead, so the per-column reads are shared-memory
         // broadcasts.  Buffer (job & 1) is rewritten only after every epilogue
@@ -423,8 +424,10 @@ __global__ void __launch_bounds__(tc_threads<NH>(), 1)
         int32_t pre1 = 0;
         auto rec_load = [&](int ctn) {
             if (MODE == MODE_SCREEN) {
-                if (te < 128) pre4 = __ldg(p.cinfo + ctn * 128 + te);
-                else if (te < 256) pre2 = __ldg(p.cinfoz + ctn * 128 + (te - 128));
+                if (te < 128) {
+                    const float4 ci = __ldg(p.cinfo + ctn * 128 + te);
+                    pre2 = make_float2(ci.x, ci.y);
+                }
             } else if (MODE == MODE_RBQ1) {
                 if (te < 128) pre4 = __ldg(p.rinfo + ctn * 128 + te);
                 else if (te < 256) pre4 = __ldg(p.rinfoq + ctn * 128 + (te - 128));
@@ -435,8 +438,7 @@ __global__ void __launch_bounds__(tc_threads<NH>(), 1)
         auto rec_store = [&](uint32_t buf) {
             uint8_t *rb = rec_base + buf * REC_BYTES;
             if (MODE == MODE_SCREEN) {
-                if (te < 128) reinterpret_cast<float4 *>(rb)[te] = pre4;
-                else if (te < 256) reinterpret_cast<float2 *>(rb + 2048)[te - 128] = pre2;
+                if (te < 128) reinterpret_cast<float2 *>(rb)[te] = pre2;
             } else if (MODE == MODE_RBQ1) {
                 if (te < 256) reinterpret_cast<float4 *>(rb)[te] = pre4;
             } else {
@@ -455,10 +457,12 @@ __global__ void __launch_bounds__(tc_threads<NH>(), 1)
             screen_init(sr);
             int32_t best = 0x7fffffff, besti = 0x7fffffff;
             float fbest = INFINITY;
-            float a2 = 0.0f, rnx2 = 0.0f, rf2 = 0.0f, rpc = 0.0f;
+            float a2 = 0.0f, w2 = 0.0f, rnx2 = 0.0f, rf2 = 0.0f, rpc = 0.0f;
             int32_t nxr = 0;
             if (MODE == MODE_SCREEN) {
                 a2 = valid ? 2.0f * p.xinfo[row].x : 0.0f;
+                // 2 W_row, W_row = 2 ||x~|| max h' + max z >= every pair's half-width
+                w2 = 2.0f * __fmaf_ru(a2, __ldg(p.hz), __ldg(p.hz + 1));
             } else if (MODE == MODE_SQ8) {
                 nxr = valid ? p.nx[row] : 0;
             } else {
@@ -487,38 +491,32 @@ __global__ void __launch_bounds__(tc_threads<NH>(), 1)
                     uint32_t v[32];
                     tmem_ld32(taddr + c * 32, v);
                     if (MODE == MODE_SCREEN) {
-                        // pass 1, two columns per packed op: m = ||c||^2 - 2 acc,
-                        // w = 2 ||x~|| h' + z; L = m - w (kept in v), U = m + w.
-                        // Records past k have ||c||^2 = +inf, so L = U = +inf.
-                        float cu[4], cl[4];
+                        // pass 1, two columns per packed op: s~ = ||c||^2 - 2 acc (kept in
+                        // v) and the chunk's smallest s~.  Records past k have ||c||^2 =
+                        // +inf, so s~ = +inf.
+                        float cm[4];
 #pragma unroll
                         for (int g = 0; g < 4; ++g) {
-                            asm volatile("" ::: "memory");  // bounds register pressure
-                            cu[g] = INFINITY;
-                            cl[g] = INFINITY;
+                            cm[g] = INFINITY;
 #pragma unroll
                             for (int i = 8 * g; i < 8 * g + 8; i += 2) {
-                                const float4 ci = reinterpret_cast<const float4 *>(rbuf)[(cc + i) >> 1];
-                                const float2 cz = reinterpret_cast<const float2 *>(rbuf + 2048)[(cc + i) >> 1];
+                                const float2 c2 = reinterpret_cast<const float2 *>(rbuf)[(cc + i) >> 1];
                                 const float2 acc = make_float2(__uint_as_float(v[i]), __uint_as_float(v[i + 1]));
-                                const float2 m = ffma2(make_float2(-2.0f, -2.0f), acc, make_float2(ci.x, ci.y));
-                                const float2 w = ffma2(make_float2(a2, a2), make_float2(ci.z, ci.w), cz);
-                                const float2 U = fadd2(m, w);
-                                const float2 L = fsub2(m, w);
-                                cu[g] = fminf(cu[g], fminf(U.x, U.y));
-                                cl[g] = fminf(cl[g], fminf(L.x, L.y));
-                                v[i] = __float_as_uint(L.x);
-                                v[i + 1] = __float_as_uint(L.y);
+                                const float2 st = ffma2(make_float2(-2.0f, -2.0f), acc, c2);
+                                cm[g] = fminf(cm[g], fminf(st.x, st.y));
+                                v[i] = __float_as_uint(st.x);
+                                v[i + 1] = __float_as_uint(st.y);
                             }
                         }
-                        sr.umin = fminf(sr.umin, fminf(fminf(cu[0], cu[1]), fminf(cu[2], cu[3])));
-                        const float lmin = fminf(fminf(cl[0], cl[1]), fminf(cl[2], cl[3]));
-                        // pass 2 (rare once Umin is small): pairs that can still be the nearest
-                        if (lmin <= sr.umin) {
+                        sr.umin = fminf(sr.umin, fminf(fminf(cm[0], cm[1]), fminf(cm[2], cm[3])));
+                        const float thr = __fadd_ru(sr.umin, w2);
+                        // pass 2 (rare once the running minimum is small): pairs within
+                        // 2 W_row of the running minimum of s~ could still be the nearest
+                        if (fminf(fminf(cm[0], cm[1]), fminf(cm[2], cm[3])) <= thr) {
                             uint32_t mask = 0;
 #pragma unroll
                             for (int i = 0; i < 32; ++i)
-                                mask |= (__uint_as_float(v[i]) <= sr.umin ? 1u : 0u) << i;
+                                mask |= (__uint_as_float(v[i]) <= thr ? 1u : 0u) << i;
                             while (mask) {
                                 const int i = __ffs(mask) - 1;
                                 mask &= mask - 1;
@@ -636,19 +634,48 @@ __global__ void __launch_bounds__(tc_threads<NH>(), 1)
                     }
                 }
                 if (MODE == MODE_SCREEN) {
+                    // The nearest centroid j* has s~_j* <= min s~ + 2 W_row (its own
+                    // and the argmin's intervals), so it is a kept candidate unless the
+                    // list overflowed (Lev inside the threshold).
+                    const float thr = __fadd_ru(sr.umin, w2);
                     int ncert = 0;
 #pragma unroll
-                    for (int t = 0; t < TCAND; ++t) ncert += (sr.L[t] <= sr.umin) ? 1 : 0;
-                    const bool overflow = !(sr.lev > sr.umin);
-                    const int first = sr.J[0] < p.k ? sr.J[0] : 0;
+                    for (int t = 0; t < TCAND; ++t) ncert += (sr.L[t] <= thr) ? 1 : 0;
+                    const bool overflow = !(sr.lev > thr);
+                    int nk = ncert;
+                    int kj[TCAND];
+#pragma unroll
+                    for (int t = 0; t < TCAND; ++t) kj[t] = sr.J[t];
+                    if (!overflow && ncert >= 2) {
+                        // refine with each candidate's own interval [s~ - w, s~ + w],
+                        // w = 2 ||x~|| h'_j + z_j (rounded outwards)
+                        float lo[TCAND], umin = INFINITY;
+#pragma unroll
+                        for (int t = 0; t < TCAND; ++t) {
+                            lo[t] = INFINITY;
+                            if (t < ncert) {
+                                const int j = sr.J[t];
+                                const float4 ci = __ldg(p.cinfo + (j >> 1));
+                                const float2 cz = __ldg(p.cinfoz + (j >> 1));
+                                const float w = __fmaf_ru(a2, (j & 1) ? ci.w : ci.z, (j & 1) ? cz.y : cz.x);
+                                umin = fminf(umin, __fadd_ru(sr.L[t], w));
+                                lo[t] = __fsub_rd(sr.L[t], w);
+                            }
+                        }
+                        nk = 0;
+#pragma unroll
+                        for (int t = 0; t < TCAND; ++t)
+                            if (t < ncert && lo[t] <= umin) kj[nk++] = sr.J[t];
+                    }
+                    const int first = kj[0] < p.k ? kj[0] : 0;
                     p.assign[row] = first;
-                    if (!overflow && ncert == 1) {
+                    if (!overflow && nk == 1) {
                         // decided by the screen
-                    } else if (!overflow && ncert >= 2) {
+                    } else if (!overflow && nk >= 2) {
                         int32_t *cr = p.cand + row * (TCAND + 1);
 #pragma unroll
-                        for (int t = 0; t < TCAND; ++t) cr[t] = sr.J[t];
-                        cr[TCAND] = ncert;
+                        for (int t = 0; t < TCAND; ++t) cr[t] = kj[t];
+                        cr[TCAND] = nk;
                         p.resc_rows[atomicAdd(&p.counters[0], 1)] = (int32_t)row;
                     } else {
                         p.fall_rows[atomicAdd(&p.counters[1], 1)] = (int32_t)row;
@@ -782,11 +809,12 @@ __global__ void screen_prep_sq8_kernel(const uint8_t *__restrict__ X, int64_t n,
 // z = eps_s ||c||^2, where rho_max >= ||x~ - x|| / ||x~|| over all points, so
 // |s~ - s| <= 2 ||x~|| h' + z = w (the half-width of the pair's interval).
 // Records j in [k, kp) get ||c||^2 = +inf so they never matter.  Layout:
-// column pair p = (2p, 2p+1) -> cinfo[p] = (||c||^2 x2, h' x2), cinfoz[p] = (z x2).
+// column pair p = (2p, 2p+1) -> cinfo[p] = (||c||^2 x2, h' x2), cinfoz[p] = (z x2);
+// hz_bits (zeroed by the caller) receives max h' and max z over j < k.
 __global__ void cprep_f32_kernel(const float *__restrict__ C, int k, int kp, int d, int dp,
                                  float eps_acc, float eps_s, const float *__restrict__ rho_max,
                                  __nv_bfloat16 *__restrict__ cs, float4 *__restrict__ cinfo,
-                                 float2 *__restrict__ cinfoz) {
+                                 float2 *__restrict__ cinfoz, unsigned int *__restrict__ hz_bits) {
     const int lane = threadIdx.x & 31;
     const int warp = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
     const int nw = (gridDim.x * blockDim.x) >> 5;
@@ -824,8 +852,12 @@ __global__ void cprep_f32_kernel(const float *__restrict__ C, int k, int kp, int
             const double h = (e + ((double)eps_acc + (double)eps_s) * g + rho * cn) * up;
             const double z = (double)eps_s * c2 * up;
             cf[4 * pp + o] = __double2float_rn(c2);
-            cf[4 * pp + 2 + o] = __double2float_ru(h);
-            zf[2 * pp + o] = __double2float_ru(z);
+            const float hf = __double2float_ru(h), zf1 = __double2float_ru(z);
+            cf[4 * pp + 2 + o] = hf;
+            zf[2 * pp + o] = zf1;
+            // maxima over the centroids (non-negative: bits order like values)
+            atomicMax(hz_bits, __float_as_uint(hf));
+            atomicMax(hz_bits + 1, __float_as_uint(zf1));
         }
     }
 }
@@ -1168,7 +1200,7 @@ int tc_screen_prep(const skm_data *x, void *screen, cudaStream_t st) {
 void tc_plan(int repr, int64_t n, int d, int k, const void *x, const void *screen, Carver &cv,
              TcAssignBufs &b) {
     b.stats = cv.take<int64_t>(4);
-    b.counters = cv.take<int32_t>(4);
+    b.counters = cv.take<int32_t>(8);  // [4], [5]: SCREEN max h', max z (float bits)
     if (repr < 0) return;  // statistics only
     const int dp = round8(d);
     const bool dense = repr == SKM_REPR_F32 || repr == SKM_REPR_BF16 ||
@@ -1220,12 +1252,14 @@ int tc_assign_float(const skm_data *x, const float *C, int k, int32_t *assign, f
     const float eps_acc = (float)((nkc * (BK / 16) + 4) * 0x1p-18);
     const float eps_s = 0x1p-21f;
     const int kp = (int)(cdiv(k, BN) * BN);
+    SKM_CUDA_TRY(cudaMemsetAsync(b.counters, 0, sizeof(int32_t) * 8, st));
     cprep_f32_kernel<<<grid_warps(kp), 256, 0, st>>>(C, k, kp, d, dp, eps_acc, eps_s, v.rho_max,
-                                                     (__nv_bfloat16 *)b.cs, b.cinfo, b.cinfoz);
+                                                     (__nv_bfloat16 *)b.cs, b.cinfo, b.cinfoz,
+                                                     reinterpret_cast<unsigned int *>(b.counters + 4));
     SKM_CUDA_TRY(launched());
-    SKM_CUDA_TRY(cudaMemsetAsync(b.counters, 0, sizeof(int32_t) * 4, st));
     TcParams p{};
     p.cinfo = b.cinfo;
+    p.hz = reinterpret_cast<const float *>(b.counters + 4);
     p.cinfoz = b.cinfoz;
     p.xinfo = v.xinfo;
     p.cand = b.cand;
