@@ -53,8 +53,13 @@ constexpr int TCAND = 4;
 constexpr unsigned long long WAIT_LIMIT_NS = 2000000000ull;  // 2 s per barrier wait
 
 enum { MODE_SCREEN = 0, MODE_SQ8 = 1, MODE_RBQ1 = 2 };
-// epilogue warps per TMEM lane quarter, by mode
+// epilogue warps per TMEM lane quarter, and CTAs per cluster (centroid
+// slices multicast across the cluster), by mode.  Clusters of 2 run
+// correctly but measured slower on GB300 (the pair's pipelines wait on each
+// other's slowest epilogue: fp32 0.999 vs 0.956 ms, 1-bit 0.602 vs 0.554 ms
+// at 1M x 1000 x 768), so every mode runs one CTA per cluster.
 constexpr int TC_NH[3] = {4, 2, 4};
+constexpr int TC_CL[3] = {1, 1, 1};
 
 // Epilogue shape: NH warps per TMEM lane quarter (column slices of 256 / NH).
 template <int NH>
@@ -155,6 +160,37 @@ __device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap *map
         "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(bar)
         : "memory");
 }
+// Multicast form: the box lands at the same shared-memory offset in every CTA
+// of the cluster named in `mask`, and each of their mbarriers at `bar`
+// receives the completed bytes.
+__device__ __forceinline__ void tma_load_2d_mc(uint32_t dst, const CUtensorMap *map, int x, int y,
+                                               uint32_t bar, uint16_t mask) {
+    asm volatile(
+        "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes.multicast::cluster"
+        " [%0], [%1, {%2, %3}], [%4], %5;" ::"r"(dst),
+        "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(bar), "h"(mask)
+        : "memory");
+}
+__device__ __forceinline__ uint32_t cluster_rank() {
+    uint32_t r;
+    asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+    return r;
+}
+__device__ __forceinline__ uint32_t cluster_index() {
+    uint32_t r;
+    asm volatile("mov.u32 %0, %%clusterid.x;" : "=r"(r));
+    return r;
+}
+__device__ __forceinline__ uint32_t cluster_count() {
+    uint32_t r;
+    asm volatile("mov.u32 %0, %%nclusterid.x;" : "=r"(r));
+    return r;
+}
+// every thread of every CTA of the cluster
+__device__ __forceinline__ void cluster_sync_all() {
+    asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" ::
+                     : "memory");
+}
 __device__ __forceinline__ void tc_fence_before() {
     asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
 }
@@ -165,6 +201,15 @@ __device__ __forceinline__ void tc_commit(uint32_t bar) {
     asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(
                      bar)
                  : "memory");
+}
+// arrive on the mbarrier at `bar` in every CTA of the cluster named in `mask`
+// once the MMAs issued so far have completed
+__device__ __forceinline__ void tc_commit_mc(uint32_t bar, uint16_t mask) {
+    asm volatile(
+        "tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64 [%0], %1;" ::"r"(
+            bar),
+        "h"(mask)
+        : "memory");
 }
 __device__ __forceinline__ void tc_mma(uint32_t dtmem, uint64_t adesc, uint64_t bdesc, uint32_t idesc,
                                        uint32_t accumulate) {
@@ -313,7 +358,7 @@ __device__ __forceinline__ void screen_insert(ScreenRow &s, float L, int j) {
     }
 }
 
-template <int MODE, int NH>
+template <int MODE, int NH, int CL>
 __global__ void __launch_bounds__(tc_threads<NH>(), 1)
     tc_assign_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                      const TcParams p) {
@@ -339,7 +384,7 @@ __global__ void __launch_bounds__(tc_threads<NH>(), 1)
     if (threadIdx.x == 0) {
         for (int s = 0; s < STAGES; ++s) {
             mbar_init(full_bar(s), 1);
-            mbar_init(empty_bar(s), 1);
+            mbar_init(empty_bar(s), CL);  // one MMA commit per CTA of the cluster
         }
         for (int b = 0; b < 2; ++b) {
             mbar_init(tfull_bar(b), 1);
@@ -360,25 +405,44 @@ __global__ void __launch_bounds__(tc_threads<NH>(), 1)
     __syncthreads();
     tc_fence_after();
     const uint32_t tmem = *tmem_slot;
+    // Cluster of CL CTAs: they walk the point tiles in lockstep (CTA r of
+    // cluster c takes point tile (c + i nclusters) CL + r) over the same
+    // centroid tiles, and each loads 256 / CL rows of every centroid slice
+    // with multicast into all of them, so a slice leaves L2 once per cluster.
+    // A stage is free again once every CTA's MMAs have read it (empty
+    // barriers count CL commits).  A tile index past the last point tile
+    // loads zeros (TMA out-of-range fill) and writes nothing.
+    const uint32_t crank = CL > 1 ? cluster_rank() : 0u;
+    const int64_t g0 = CL > 1 ? (int64_t)cluster_index() : (int64_t)blockIdx.x;
+    const int64_t gstep = CL > 1 ? (int64_t)cluster_count() : (int64_t)gridDim.x;
+    const int64_t ngroups = (p.nrt + CL - 1) / CL;
+    if (CL > 1) cluster_sync_all();  // peers' barriers are initialised before any multicast
 
     if (warp == 0) {
         if (lane == 0) {  // ---------------------------------------- TMA producer
             uint32_t it = 0;
-            for (int64_t rt = blockIdx.x; rt < p.nrt; rt += gridDim.x)
+            for (int64_t g = g0; g < ngroups; g += gstep) {
+                const int64_t rt = g * CL + crank;
                 for (int ct = 0; ct < p.nct; ++ct)
                     for (int kc = 0; kc < p.nkc; ++kc, ++it) {
                         const uint32_t s = it % STAGES, ph = (it / STAGES) & 1u;
                         if (!mbar_wait(empty_bar(s), ph ^ 1u, abort_flag)) goto producer_done;
                         mbar_expect_tx(full_bar(s), A_STAGE + B_STAGE);
                         tma_load_2d(sA + s * A_STAGE, &tmA, kc * KC_ELEMS, (int)(rt * BM), full_bar(s));
-                        tma_load_2d(sB + s * B_STAGE, &tmB, kc * KC_ELEMS, ct * BN, full_bar(s));
+                        if (CL == 1)
+                            tma_load_2d(sB + s * B_STAGE, &tmB, kc * KC_ELEMS, ct * BN, full_bar(s));
+                        else
+                            tma_load_2d_mc(sB + s * B_STAGE + crank * (B_STAGE / CL), &tmB, kc * KC_ELEMS,
+                                           ct * BN + (int)crank * (BN / CL), full_bar(s),
+                                           (uint16_t)((1u << CL) - 1u));
                     }
+            }
         producer_done:;
         }
     } else if (warp == 1) {
         if (lane == 0) {  // ---------------------------------------- MMA issuer
             uint32_t it = 0, job = 0;
-            for (int64_t rt = blockIdx.x; rt < p.nrt; rt += gridDim.x)
+            for (int64_t g = g0; g < ngroups; g += gstep)
                 for (int ct = 0; ct < p.nct; ++ct, ++job) {
                     const uint32_t b = job & 1u, bph = (job >> 1) & 1u;
                     if (!mbar_wait(tempty_bar(b), bph ^ 1u, abort_flag)) goto mma_done;
@@ -397,7 +461,10 @@ __global__ void __launch_bounds__(tc_threads<NH>(), 1)
                             else
                                 tc_mma(dcol, ad + 2u * kk, bd + 2u * kk, IDESC, (kc | kk) != 0);
                         }
-                        tc_commit(empty_bar(s));
+                        if (CL == 1)
+                            tc_commit(empty_bar(s));
+                        else
+                            tc_commit_mc(empty_bar(s), (uint16_t)((1u << CL) - 1u));
                     }
                     tc_commit(tfull_bar(b));
                 }
@@ -450,7 +517,8 @@ __global__ void __launch_bounds__(tc_threads<NH>(), 1)
         // in the named barriers, so the other epilogue warps never wait on it.
         bool dead = false;
         uint32_t job = 0;
-        for (int64_t rt = blockIdx.x; rt < p.nrt; rt += gridDim.x) {
+        for (int64_t g = g0; g < ngroups; g += gstep) {
+            const int64_t rt = g * CL + crank;
             const int64_t row = rt * BM + rin;
             const bool valid = row < p.n;
             ScreenRow sr;
@@ -692,6 +760,9 @@ __global__ void __launch_bounds__(tc_threads<NH>(), 1)
     }
     tc_fence_before();
     __syncthreads();
+    // no CTA leaves while a peer may still multicast into its shared memory
+    // or arrive on its barriers
+    if (CL > 1) cluster_sync_all();
     if (warp == 1) {
         __syncwarp();
         tc_fence_after();
@@ -1059,28 +1130,67 @@ template <int MODE>
 int launch_tc(const void *xs, int64_t n, int dp, int d, const void *cs, int k, const TcParams &p0,
               cudaStream_t st) {
     constexpr int NH = TC_NH[MODE];
+    constexpr int CL = TC_CL[MODE];
     constexpr size_t SMEM = tc_smem_bytes<MODE, NH>();
     static_assert(SMEM <= 227 * 1024, "shared memory per CTA");
-    static std::once_flag attr_once[3];
-    static cudaError_t attr_err[3] = {cudaSuccess, cudaSuccess, cudaSuccess};
-    std::call_once(attr_once[MODE], [] {
-        attr_err[MODE] = cudaFuncSetAttribute(tc_assign_kernel<MODE, NH>,
-                                              cudaFuncAttributeMaxDynamicSharedMemorySize, (int)SMEM);
-    });
-    if (attr_err[MODE] != cudaSuccess)
-        return set_error(SKM_ERR_CUDA, "cudaFuncSetAttribute: %s", cudaGetErrorString(attr_err[MODE]));
+    auto kern = tc_assign_kernel<MODE, NH, CL>;
+    // per device: the attribute and the number of clusters that fit at once
+    constexpr int MAXDEV = 64;
+    static std::mutex mu;
+    static int cached_clusters[3][MAXDEV] = {};
+    int dev = 0;
+    SKM_CUDA_TRY(cudaGetDevice(&dev));
+    int max_clusters = 0;
+    {
+        std::lock_guard<std::mutex> lock(mu);
+        if (dev < MAXDEV) max_clusters = cached_clusters[MODE][dev];
+        if (max_clusters == 0) {
+            SKM_CUDA_TRY(cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)SMEM));
+            if (CL > 1) {
+                cudaLaunchConfig_t qc = {};
+                qc.gridDim = dim3((unsigned)(CL * device_sms()));
+                qc.blockDim = dim3(tc_threads<NH>());
+                qc.dynamicSmemBytes = SMEM;
+                cudaLaunchAttribute qa[1];
+                qa[0].id = cudaLaunchAttributeClusterDimension;
+                qa[0].val.clusterDim.x = CL;
+                qa[0].val.clusterDim.y = 1;
+                qa[0].val.clusterDim.z = 1;
+                qc.attrs = qa;
+                qc.numAttrs = 1;
+                SKM_CUDA_TRY(cudaOccupancyMaxActiveClusters(&max_clusters, kern, &qc));
+            } else {
+                max_clusters = device_sms();
+            }
+            if (max_clusters < 1) return set_error(SKM_ERR_CUDA, "no cluster of %d CTAs fits on this device", CL);
+            if (dev < MAXDEV) cached_clusters[MODE][dev] = max_clusters;
+        }
+    }
     CUtensorMap ma, mb;
     const int eb = MODE == MODE_RBQ1 ? 1 : 2;
     SKM_TRY(make_map(&ma, xs, n, d, dp, BM, eb));
-    SKM_TRY(make_map(&mb, cs, k, d, dp, BN, eb));
+    SKM_TRY(make_map(&mb, cs, k, d, dp, BN / CL, eb));
     TcParams p = p0;
     p.n = n;
     p.nrt = cdiv(n, BM);
     p.k = k;
     p.nct = (int)cdiv(k, BN);
     p.nkc = (int)cdiv(d, 128 / eb);
-    const int grid = (int)std::min<int64_t>(device_sms(), p.nrt);
-    tc_assign_kernel<MODE, NH><<<grid, tc_threads<NH>(), SMEM, st>>>(ma, mb, p);
+    const int64_t groups = cdiv(p.nrt, CL);
+    const int grid = CL * (int)std::min<int64_t>(max_clusters, groups);
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3((unsigned)grid);
+    cfg.blockDim = dim3(tc_threads<NH>());
+    cfg.dynamicSmemBytes = SMEM;
+    cfg.stream = st;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = CL;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    SKM_CUDA_TRY(cudaLaunchKernelEx(&cfg, kern, ma, mb, p));
     SKM_CUDA_TRY(launched());
     return SKM_OK;
 }
