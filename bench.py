@@ -489,6 +489,10 @@ def run_case(args):
         q = skm.skm_quantize(skm.REPR_SQ8, X)
         pts = skm.Points(skm.REPR_SQ8, q["codes"], d).with_screen()
         C = q["codes"][:k].clone()
+    elif args.case == "assign_prune":  # bf16 points, exact prefix-block pruning
+        Xb = X.to(torch.bfloat16).view(torch.int16).contiguous()
+        pts = skm.Points(skm.REPR_BF16, Xb, d, flags=skm.FLAG_PRUNE)
+        C = (Xb[synth.forgy_indices(n, k, seed=0).cuda()].to(torch.int32) << 16).view(torch.float32).contiguous()
     else:
         raise SystemExit(f"unknown case {args.case}")
     wsA = skm.workspace(skm.OP_ASSIGN, pts, k)
@@ -516,6 +520,102 @@ def run_case(args):
     print(json.dumps(out))
 
 
+def run_config(args):
+    """One JSON line per representation of a workload configuration: the
+    median over Lloyd iterations 2..iters of (centroid prep + assign + update)
+    timed with CUDA events, distances/s = n k / t_iter, and the assignment
+    against its roofline (2 n k d flop on the bf16 / e4m3 tensor peak)."""
+    import numpy as np
+    import torch
+
+    import paper_2608_14648_gb300 as skm
+    import synth
+
+    torch.cuda.set_device(0)
+    dev = torch.device("cuda", 0)
+    peaks = load_peaks()
+    iters = args.iters
+    name = {"c0": "tiny_f32", "c1": "emb1m_d768", "c2": "emb1m_d1024_sq8", "c3": "emb10m_d1024_rbq1",
+            "c4": "emb10m_pca256"}[args.config]
+    spec = synth.WORKLOADS[name]
+    n, k = spec.n, spec.k
+    idx = synth.forgy_indices(n, k, seed=0).to(dev)
+    X = synth.workload_points(spec, seed=0, device=dev)
+    runs = []  # (label, Points, C0, d, peak TFLOP/s, flop kind)
+    bf16_peak = peaks["bf16_tflops"]
+    if args.config in ("c0", "c1"):
+        runs.append(("fp32", skm.Points(skm.REPR_F32, X, spec.d).with_screen(), X[idx].clone(), spec.d,
+                     bf16_peak, "bf16"))
+    if args.config == "c1":
+        q = skm.skm_quantize(skm.REPR_RBQ1, X)
+        pR = skm.rbq1_points(q, spec.d).with_screen()
+        CR, _, _, _, _ = skm.skm_fit(pR, k, 0, init_idx=idx, want_objective=False, want_dist=False)
+        runs.append(("rbq1", pR, CR, spec.d, 2 * bf16_peak, "e4m3"))
+    if args.config == "c2":
+        q = skm.skm_quantize(skm.REPR_SQ8, X)
+        del X
+        runs.append(("sq8", skm.Points(skm.REPR_SQ8, q["codes"], spec.d).with_screen(),
+                     q["codes"][idx].clone(), spec.d, bf16_peak, "bf16"))
+    if args.config == "c3":
+        P = synth.haar_rotation(spec.d, 99).to(torch.float32).contiguous().to(dev)
+        Y = skm.skm_project(X, P)
+        del X
+        q = skm.skm_quantize(skm.REPR_RBQ1, Y)
+        del Y
+        pR = skm.rbq1_points(q, spec.d).with_screen()
+        CR, _, _, _, _ = skm.skm_fit(pR, k, 0, init_idx=idx, want_objective=False, want_dist=False)
+        runs.append(("rbq1", pR, CR, spec.d, 2 * bf16_peak, "e4m3"))
+    if args.config == "c4":
+        dp = 256
+        mean, P, _ = skm.skm_pca_fit(X, dp)
+        Yb = skm.skm_project(X, P, mean, out_dtype=skm.DTYPE_BF16).view(torch.int16)
+        del X
+        Cb = (Yb[idx].to(torch.int32) << 16).view(torch.float32).contiguous()
+        runs.append(("bf16_screen", skm.Points(skm.REPR_BF16, Yb, dp).with_screen(), Cb, dp, bf16_peak, "bf16"))
+        runs.append(("bf16_prune", skm.Points(skm.REPR_BF16, Yb, dp, flags=skm.FLAG_PRUNE), Cb.clone(), dp,
+                     None, "fp32 CUDA cores"))
+    torch.cuda.synchronize()
+    for label, pts, C, d, peak, kind in runs:
+        C = C.clone()
+        wsA = skm.workspace(skm.OP_ASSIGN, pts, k)
+        wsU = skm.workspace(skm.OP_UPDATE, pts, k)
+        a = torch.empty(n, dtype=torch.int32, device=dev)
+        prev = None
+        cnt = torch.zeros(k, dtype=torch.int64, device=dev)
+        stream = torch.cuda.current_stream()
+        ta, tu = [], []
+        for it in range(iters):
+            e0, e1, e2 = (torch.cuda.Event(enable_timing=True) for _ in range(3))
+            e0.record(stream)
+            skm.skm_assign(pts, C, k, prev_assign=prev, want_dist=False, ws=wsA, out=a)
+            e1.record(stream)
+            skm.skm_update(pts, a, C, counts=cnt, ws=wsU)
+            e2.record(stream)
+            torch.cuda.synchronize()
+            ta.append(e0.elapsed_time(e1))
+            tu.append(e1.elapsed_time(e2))
+            if label == "bf16_prune":
+                prev = a.clone()
+        sel = slice(1, None) if iters > 1 else slice(0, None)
+        t_a = float(np.median(ta[sel]))
+        t_u = float(np.median(tu[sel]))
+        t_it = float(np.median([x + y for x, y in zip(ta[sel], tu[sel])]))
+        out = {"config": args.config, "workload": name, "repr": label, "n": n, "d": d, "k": k,
+               "iters": iters, "ms_per_iter": round(t_it, 4), "assign_ms": round(t_a, 4),
+               "update_ms": round(t_u, 4), "distances_per_s": n * k / (t_it / 1e3)}
+        if peak:
+            ach = 2.0 * n * k * d / (t_a / 1e3) / 1e12
+            out["assign_roofline"] = {"bound": "tensor", "achieved_tflops": round(ach, 2),
+                                      "peak_tflops": peak, "frac": round(ach / peak, 4), "flop": kind}
+        if label == "bf16_prune":
+            _, _, _, _, st = skm.skm_fit(pts, k, 1, C_init=C, want_objective=False, want_dist=False)
+            out["prune_stats_2_assigns"] = st
+            out["dense_equiv_tensor_ms"] = round(2.0 * n * k * d / (bf16_peak * 1e12) * 1e3, 3)
+        print(json.dumps(out), flush=True)
+        del wsA, wsU
+        torch.cuda.empty_cache()
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -526,15 +626,21 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-popcount", action="store_true")
     ap.add_argument("--case", default=None,
-                    help="single-operation run for profiling: assign_f32|assign_rbq1|assign_sq8|update_f32|"
-                         "update_rbq1|update_sq8")
+                    help="single-operation run for profiling: assign_f32|assign_rbq1|assign_sq8|"
+                         "assign_rbq1_popcount|assign_prune|update_f32|update_rbq1|update_sq8")
     ap.add_argument("--n", type=int, default=200_000)
     ap.add_argument("--d", type=int, default=768)
     ap.add_argument("--k", type=int, default=1000)
     ap.add_argument("--reps", type=int, default=3)
+    ap.add_argument("--config", default=None, choices=["c0", "c1", "c2", "c3", "c4"],
+                    help="per-configuration Lloyd iteration timing (median of iterations 2..iters)")
+    ap.add_argument("--iters", type=int, default=10)
     args = ap.parse_args()
     if args.case:
         run_case(args)
+        return
+    if args.config:
+        run_config(args)
         return
     if args.warmup < 3:
         print("warning: fewer than 3 warm-up steps", file=sys.stderr)

@@ -1,5 +1,6 @@
-// Streamed segmented sums for the centroid update (Section 2.3 STEP 3; for
-// 1-bit codes the fused decode-average of Section 3.1 "RabitQ").
+// Streamed segmented sums for the centroid update (Section 2.3 STEP 3; SQ8
+// codes summed exactly in the code domain and, for 1-bit codes, the fused
+// decode-average of Section 3.1 "RabitQ").
 //
 // The cluster-sorted member order is cut into runs of RS_ROWS positions and
 // each of the RS_CW consumer warps of a CTA owns one run.  A producer warp
@@ -370,6 +371,93 @@ __global__ void __launch_bounds__(RS_THREADS) ring_sum_rbq1_kernel(
     ring_run(reinterpret_cast<const uint8_t *>(codes), perm, nval, L, flag, cons);
 }
 
+// --------------------------------------------------------------- SQ8 rows
+// S[c][i] += code_i (int64).  Lane l holds the 16-byte column groups
+// l + 32 t (t < NG).  Inside a run (at most RS_ROWS rows between flushes)
+// each 32-bit word's four codes are summed as two words of two 16-bit lanes
+// (bytes 0, 2 and bytes 1, 3), which cannot overflow (128 x 255 < 2^16).
+template <int NG>
+struct Sq8Cons {
+    const int32_t *scl;
+    unsigned long long *S;
+    int d;
+    uint32_t ev[4 * NG], od[4 * NG];  // per word: bytes 0,2 and bytes 1,3
+    int cur;
+    int64_t q0;
+    int clw, cln;
+    int cnt;
+    __device__ __forceinline__ void flush(int c, int lane) {
+#pragma unroll
+        for (int t = 0; t < NG; ++t)
+#pragma unroll
+            for (int u = 0; u < 4; ++u) {
+                const int col = 16 * (lane + 32 * t) + 4 * u;
+                if (col < d) {
+                    unsigned long long *dst = S + (int64_t)c * d + col;
+                    const uint32_t e = ev[4 * t + u], o = od[4 * t + u];
+                    if (e & 0xffffu) atomicAdd(dst + 0, (unsigned long long)(e & 0xffffu));
+                    if (o & 0xffffu) atomicAdd(dst + 1, (unsigned long long)(o & 0xffffu));
+                    if (e >> 16) atomicAdd(dst + 2, (unsigned long long)(e >> 16));
+                    if (o >> 16) atomicAdd(dst + 3, (unsigned long long)(o >> 16));
+                }
+                ev[4 * t + u] = 0u;
+                od[4 * t + u] = 0u;
+            }
+    }
+    __device__ __forceinline__ void start(int64_t q0_, int cnt_, int lane) {
+        q0 = q0_;
+        cnt = cnt_;
+#pragma unroll
+        for (int t = 0; t < 4 * NG; ++t) ev[t] = od[t] = 0u;
+        clw = lane < cnt ? __ldg(scl + q0 + lane) : -1;
+        cln = 32 + lane < cnt ? __ldg(scl + q0 + 32 + lane) : -1;
+        cur = __shfl_sync(0xffffffffu, clw, 0);
+    }
+    __device__ __forceinline__ void row(int i, const uint8_t *slot, int lane) {
+        if ((i & 31) == 0 && i > 0) {
+            clw = cln;
+            const int nx = i + 32 + lane;
+            cln = nx < cnt ? __ldg(scl + q0 + nx) : -1;
+        }
+        const int c = __shfl_sync(0xffffffffu, clw, i & 31);
+        if (c != cur) {
+            flush(cur, lane);
+            cur = c;
+        }
+        const int ng16 = d >> 4;  // 16-byte groups (d % 16 == 0 on this path)
+#pragma unroll
+        for (int t = 0; t < NG; ++t) {
+            const int gidx = lane + 32 * t;
+            if (gidx < ng16) {
+                const uint4 w = reinterpret_cast<const uint4 *>(slot)[gidx];
+                ev[4 * t + 0] += w.x & 0x00ff00ffu;
+                od[4 * t + 0] += (w.x >> 8) & 0x00ff00ffu;
+                ev[4 * t + 1] += w.y & 0x00ff00ffu;
+                od[4 * t + 1] += (w.y >> 8) & 0x00ff00ffu;
+                ev[4 * t + 2] += w.z & 0x00ff00ffu;
+                od[4 * t + 2] += (w.z >> 8) & 0x00ff00ffu;
+                ev[4 * t + 3] += w.w & 0x00ff00ffu;
+                od[4 * t + 3] += (w.w >> 8) & 0x00ff00ffu;
+            }
+        }
+    }
+    __device__ __forceinline__ void finish(int lane) { flush(cur, lane); }
+};
+
+template <int NG>
+__global__ void __launch_bounds__(RS_THREADS) ring_sum_sq8_kernel(
+    const uint8_t *__restrict__ codes, int d, const int32_t *__restrict__ perm,
+    const int32_t *__restrict__ scl, const int64_t *__restrict__ offsets, int k,
+    unsigned long long *__restrict__ S, RingLayout L, int32_t *flag) {
+    const int64_t nval = offsets[k];
+    if ((int64_t)blockIdx.x * RS_CW * RS_ROWS >= nval) return;
+    Sq8Cons<NG> cons;
+    cons.scl = scl;
+    cons.S = S;
+    cons.d = d;
+    ring_run(codes, perm, nval, L, flag, cons);
+}
+
 bool ring_layout(uint32_t rb, RingLayout &L) {
     if (rb == 0 || rb % 16 != 0) return false;
     L.rb = (int)rb;
@@ -439,6 +527,38 @@ cudaError_t launch_ring_sum_float(const void *X, int x_is_bf16, int64_t n, int d
                          : launch_float_nf<false, double>(nf, X, n, d, perm, scl, offsets, k, S_d, L, flag, st);
     return x_is_bf16 ? launch_float_nf<true, float>(nf, X, n, d, perm, scl, offsets, k, S_f, L, flag, st)
                      : launch_float_nf<false, float>(nf, X, n, d, perm, scl, offsets, k, S_f, L, flag, st);
+}
+
+bool ring_sum_sq8_ok(const void *codes, int d) {
+    RingLayout L;
+    return d % 16 == 0 && d <= 4096 && (reinterpret_cast<uintptr_t>(codes) & 15u) == 0 &&
+           ring_layout((uint32_t)d, L);
+}
+
+cudaError_t launch_ring_sum_sq8(const uint8_t *codes, int64_t n, int d, const int32_t *perm,
+                                const int32_t *scl, const int64_t *offsets, int k, int64_t *S,
+                                int32_t *flag, cudaStream_t st) {
+    if (n == 0) return cudaSuccess;
+    RingLayout L;
+    if (!ring_layout((uint32_t)d, L)) return cudaErrorInvalidValue;
+    const size_t smem = L.bytes();
+    const unsigned g = ring_blocks(n);
+    auto S64 = reinterpret_cast<unsigned long long *>(S);
+    const int q = (d / 16 + 31) / 32;  // 16-byte groups per lane
+#define RS_CASE(NGV)                                                                                \
+    if (q <= NGV) {                                                                                 \
+        auto kern = ring_sum_sq8_kernel<NGV>;                                                       \
+        cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem); \
+        if (e != cudaSuccess) return e;                                                             \
+        kern<<<g, RS_THREADS, smem, st>>>(codes, d, perm, scl, offsets, k, S64, L, flag);            \
+        return launched();                                                                          \
+    }
+    RS_CASE(1)
+    RS_CASE(2)
+    RS_CASE(4)
+    RS_CASE(8)
+#undef RS_CASE
+    return cudaErrorInvalidValue;
 }
 
 cudaError_t launch_ring_sum_rbq1(const uint32_t *codes, const int64_t *fqs, int64_t n, int d,

@@ -117,7 +117,7 @@ struct UpdateBufs {
     int64_t *offsets = nullptr;
     int64_t *fq = nullptr;    // RBQ1: fixed-point weights round(F 2^e)
     float *sumf = nullptr;    // F32/BF16: cluster sums [k][d]
-    int64_t *sumi = nullptr;  // RBQ1: cluster sums [k][d + 1]
+    int64_t *sumi = nullptr;  // RBQ1: cluster sums [k][d + 1]; SQ8: [k][d]
     int32_t *flag = nullptr;  // raised by a streamed-sum wait that gave up
 };
 
@@ -131,6 +131,7 @@ static void plan_update(const skm_data *x, int k, Carver &cv, UpdateBufs &b) {
         b.fq = cv.take<int64_t>(x->n);
         b.sumi = cv.take<int64_t>((size_t)k * (x->d + 1));
     }
+    if (x->repr == SKM_REPR_SQ8) b.sumi = cv.take<int64_t>((size_t)k * x->d);
     if (x->repr == SKM_REPR_F32 || x->repr == SKM_REPR_BF16) b.sumf = cv.take<float>((size_t)k * x->d);
     b.flag = cv.take<int32_t>(1);
 }
@@ -239,11 +240,20 @@ static int do_update(const skm_data *x, const int32_t *assign, int k, void *C, i
             SKM_CUDA_TRY(launch_finalize_float32(b.sumf, counts, k, d, static_cast<float *>(C), st));
         break;
     }
-    case SKM_REPR_SQ8:
-        SKM_CUDA_TRY(launch_segsum_sq8(static_cast<const uint8_t *>(x->x), d, b.perm, b.offsets, k,
-                                       static_cast<uint8_t *>(C), static_cast<int64_t *>(partial),
-                                       st));
+    case SKM_REPR_SQ8: {
+        const uint8_t *codes = static_cast<const uint8_t *>(x->x);
+        if (ring_sum_sq8_ok(codes, d)) {
+            int64_t *S = partial ? static_cast<int64_t *>(partial) : b.sumi;
+            if (!partial) SKM_CUDA_TRY(cudaMemsetAsync(S, 0, sizeof(int64_t) * (size_t)k * d, st));
+            SKM_CUDA_TRY(launch_ring_sum_sq8(codes, n, d, b.perm, b.scl, b.offsets, k, S, b.flag, st));
+            if (!partial)
+                SKM_CUDA_TRY(launch_finalize_sq8(S, counts, k, d, static_cast<uint8_t *>(C), st));
+        } else {
+            SKM_CUDA_TRY(launch_segsum_sq8(codes, d, b.perm, b.offsets, k, static_cast<uint8_t *>(C),
+                                           static_cast<int64_t *>(partial), st));
+        }
         break;
+    }
     case SKM_REPR_RBQ1: {
         SKM_CUDA_TRY(launch_rbq1_fq(x->F, b.perm, b.offsets, k, n, e, b.fq, st));
         int64_t *T = partial ? static_cast<int64_t *>(partial) : b.sumi;

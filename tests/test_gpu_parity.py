@@ -110,7 +110,8 @@ def _skewed_assign(n, k, seed):
 
 @pytest.mark.parametrize("repr_name,n,d,k", [("f32", 70001, 128, 500), ("f32", 9000, 1536, 40),
                                              ("bf16", 20011, 1024, 300), ("rbq1", 70001, 128, 500),
-                                             ("rbq1", 20011, 1024, 300)])
+                                             ("rbq1", 20011, 1024, 300), ("sq8", 70001, 128, 500),
+                                             ("sq8", 20011, 1024, 300), ("sq8", 5003, 48, 20)])
 def test_update_skewed_clusters(skm, repr_name, n, d, k):
     """Runs of the sorted order that cross many small clusters and one giant
     cluster shared by hundreds of runs; ragged last run; skipped points."""
@@ -118,6 +119,16 @@ def test_update_skewed_clusters(skm, repr_name, n, d, k):
     a = _skewed_assign(n, k, seed=d)
     ok = (a >= 0).numpy()
     C0 = X[:k].clone()
+    if repr_name == "sq8":
+        q = skm.skm_quantize(skm.REPR_SQ8, X.to(DEV))
+        pts = skm.Points(skm.REPR_SQ8, q["codes"], d)
+        codes = q["codes"].cpu().numpy()
+        Cc = q["codes"][:k].clone()
+        Cn, counts = skm.skm_update(pts, a.to(DEV), Cc.clone())
+        Co, co = oracle.update_sq8(codes[ok], a.numpy()[ok], Cc.cpu().numpy())
+        np.testing.assert_array_equal(counts.cpu().numpy(), co)
+        np.testing.assert_array_equal(Cn.cpu().numpy(), Co)
+        return
     if repr_name == "rbq1":
         r = skm.skm_quantize(skm.REPR_RBQ1, X.to(DEV))
         pts = skm.rbq1_points(r, d)
