@@ -32,7 +32,13 @@ __device__ __forceinline__ void argmin_merge(float &bd, int &bi, float d, int i)
 
 // rows == nullptr: rows 0..nrows-1.  Otherwise the rows are rows[0..count)
 // with count = *nrows_dev (a device-side list, e.g. the rows a screen could
-// not decide).  Blocks stride over 64-row tiles.
+// not decide).  Blocks stride over work items of 64 rows.  With `keys` (one
+// per listed row, preset to ~0) the centroids are also split across the grid
+// when the list is short (a handful of rows against thousands of centroids
+// would otherwise run on a few SMs): each work item covers a range of
+// centroid tiles and merges (dist bits << 32 | index) into its rows' keys with
+// atomicMin — non-negative distances order like their bit patterns, so the
+// smallest key is the nearest centroid with ties to the lowest index.
 template <typename TX>
 __global__ void __launch_bounds__(256) assign_exact_kernel(const TX *__restrict__ X,
                                                            const int32_t *__restrict__ rows,
@@ -40,13 +46,23 @@ __global__ void __launch_bounds__(256) assign_exact_kernel(const TX *__restrict_
                                                            int64_t nrows_arg, int d,
                                                            const float *__restrict__ C, int k,
                                                            int32_t *__restrict__ assign,
-                                                           float *__restrict__ dist) {
+                                                           float *__restrict__ dist,
+                                                           unsigned long long *__restrict__ keys) {
     __shared__ __align__(16) float xs[32][68];
     __shared__ __align__(16) float cs[32][68];
     const int tid = threadIdx.x;
     const int ty = tid >> 4, tx = tid & 15;
     const int64_t nrows = nrows_dev ? (int64_t)*nrows_dev : nrows_arg;
-    for (int64_t row0 = (int64_t)blockIdx.x * 64; row0 < nrows; row0 += (int64_t)gridDim.x * 64) {
+    const int64_t rtiles = (nrows + 63) / 64;
+    const int ktiles = (k + 63) / 64;
+    int nsplit = 1;
+    if (keys && rtiles > 0) nsplit = (int)max((int64_t)1, min((int64_t)ktiles, (int64_t)gridDim.x / rtiles));
+    const int tps = (ktiles + nsplit - 1) / nsplit;  // centroid tiles per split
+    const int64_t nwork = rtiles * nsplit;
+    for (int64_t w = blockIdx.x; w < nwork; w += gridDim.x) {
+        const int64_t row0 = (w / nsplit) * 64;
+        const int cbeg = (int)(w % nsplit) * tps * 64;
+        const int cend = min(k, cbeg + tps * 64);
         __syncthreads();
 
         // the point rows this block owns (indirect when `rows` is given)
@@ -77,7 +93,7 @@ __global__ void __launch_bounds__(256) assign_exact_kernel(const TX *__restrict_
             besti[i] = 0x7fffffff;
         }
 
-        for (int c0 = 0; c0 < k; c0 += 64) {
+        for (int c0 = cbeg; c0 < cend; c0 += 64) {
             float acc[4][4];
 #pragma unroll
             for (int i = 0; i < 4; ++i)
@@ -93,7 +109,7 @@ __global__ void __launch_bounds__(256) assign_exact_kernel(const TX *__restrict_
                     float xv = 0.0f, cv = 0.0f;
                     if (dim < d) {
                         if (lval[q]) xv = load_x<TX>(X + lrow[q] * d + dim);
-                        if (c0 + r < k) cv = __ldg(C + (int64_t)(c0 + r) * d + dim);
+                        if (c0 + r < cend) cv = __ldg(C + (int64_t)(c0 + r) * d + dim);
                     }
                     xs[ld][r] = xv;
                     cs[ld][r] = cv;
@@ -122,7 +138,7 @@ __global__ void __launch_bounds__(256) assign_exact_kernel(const TX *__restrict_
 #pragma unroll
                 for (int j = 0; j < 4; ++j) {
                     const int cj = c0 + tx * 4 + j;
-                    if (cj < k) argmin_merge(bd, bi, acc[i][j], cj);
+                    if (cj < cend) argmin_merge(bd, bi, acc[i][j], cj);
                 }
 #pragma unroll
                 for (int o = 8; o > 0; o >>= 1) {
@@ -137,11 +153,35 @@ __global__ void __launch_bounds__(256) assign_exact_kernel(const TX *__restrict_
 #pragma unroll
             for (int i = 0; i < 4; ++i)
                 if (pval[i]) {
-                    assign[prow[i]] = besti[i];
-                    if (dist) dist[prow[i]] = best[i];
+                    if (keys) {
+                        if (besti[i] != 0x7fffffff)
+                            atomicMin(keys + row0 + ty * 4 + i,
+                                      ((unsigned long long)__float_as_uint(best[i]) << 32) | (uint32_t)besti[i]);
+                    } else {
+                        assign[prow[i]] = besti[i];
+                        if (dist) dist[prow[i]] = best[i];
+                    }
                 }
         }
-    }  // row tiles
+    }  // work items
+}
+
+__global__ void keys_init_kernel(const int32_t *__restrict__ count, unsigned long long *__restrict__ keys) {
+    const int64_t c = *count;
+    for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < c; i += (int64_t)gridDim.x * blockDim.x)
+        keys[i] = ~0ull;
+}
+
+__global__ void keys_finish_kernel(const int32_t *__restrict__ rows, const int32_t *__restrict__ count,
+                                   const unsigned long long *__restrict__ keys, int32_t *__restrict__ assign,
+                                   float *__restrict__ dist) {
+    const int64_t c = *count;
+    for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < c; i += (int64_t)gridDim.x * blockDim.x) {
+        const unsigned long long key = keys[i];
+        if (key == ~0ull) continue;  // no centroid (k == 0 cannot happen on this path)
+        assign[rows[i]] = (int32_t)(key & 0xffffffffull);
+        if (dist) dist[rows[i]] = __uint_as_float((uint32_t)(key >> 32));
+    }
 }
 
 static unsigned blocks_for_rows(int64_t nrows) {
@@ -154,7 +194,7 @@ cudaError_t launch_assign_exact_f32(const float *X, int64_t n, int d, const floa
                                     int32_t *assign, float *dist, cudaStream_t st) {
     if (n == 0) return cudaSuccess;
     assign_exact_kernel<float><<<blocks_for_rows(n), 256, 0, st>>>(X, nullptr, nullptr, n, d, C,
-                                                                   k, assign, dist);
+                                                                   k, assign, dist, nullptr);
     return launched();
 }
 
@@ -162,22 +202,31 @@ cudaError_t launch_assign_exact_bf16(const uint16_t *X, int64_t n, int d, const 
                                      int32_t *assign, float *dist, cudaStream_t st) {
     if (n == 0) return cudaSuccess;
     assign_exact_kernel<uint16_t><<<blocks_for_rows(n), 256, 0, st>>>(X, nullptr, nullptr, n, d,
-                                                                      C, k, assign, dist);
+                                                                      C, k, assign, dist, nullptr);
     return launched();
 }
 
 cudaError_t launch_assign_exact_rows(const void *X, int x_is_bf16, const int32_t *rows,
                                      const int32_t *count_dev, int64_t max_rows, int d,
                                      const float *C, int k, int32_t *assign, float *dist,
-                                     cudaStream_t st) {
+                                     unsigned long long *keys, cudaStream_t st) {
     if (max_rows == 0) return cudaSuccess;
-    const unsigned g = blocks_for_rows(max_rows);
+    // enough blocks to split the centroids when only a few rows are listed
+    const unsigned g = keys ? 152u * 4u : blocks_for_rows(max_rows);
+    if (keys) {
+        keys_init_kernel<<<152, 256, 0, st>>>(count_dev, keys);
+        cudaError_t e = launched();
+        if (e != cudaSuccess) return e;
+    }
     if (x_is_bf16)
         assign_exact_kernel<uint16_t><<<g, 256, 0, st>>>(static_cast<const uint16_t *>(X), rows,
-                                                         count_dev, 0, d, C, k, assign, dist);
+                                                         count_dev, 0, d, C, k, assign, dist, keys);
     else
         assign_exact_kernel<float><<<g, 256, 0, st>>>(static_cast<const float *>(X), rows,
-                                                      count_dev, 0, d, C, k, assign, dist);
+                                                      count_dev, 0, d, C, k, assign, dist, keys);
+    cudaError_t e = launched();
+    if (e != cudaSuccess || !keys) return e;
+    keys_finish_kernel<<<152, 256, 0, st>>>(rows, count_dev, keys, assign, dist);
     return launched();
 }
 

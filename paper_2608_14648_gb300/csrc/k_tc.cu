@@ -581,10 +581,16 @@ __global__ void __launch_bounds__(tc_threads<NH>(), 1)
                         // pass 2 (rare once the running minimum is small): pairs within
                         // 2 W_row of the running minimum of s~ could still be the nearest
                         if (fminf(fminf(cm[0], cm[1]), fminf(cm[2], cm[3])) <= thr) {
+                            // only the 8-column groups whose minimum is inside
                             uint32_t mask = 0;
 #pragma unroll
-                            for (int i = 0; i < 32; ++i)
-                                mask |= (__uint_as_float(v[i]) <= thr ? 1u : 0u) << i;
+                            for (int g = 0; g < 4; ++g) {
+                                if (cm[g] <= thr) {
+#pragma unroll
+                                    for (int i = 8 * g; i < 8 * g + 8; ++i)
+                                        mask |= (__uint_as_float(v[i]) <= thr ? 1u : 0u) << i;
+                                }
+                            }
                             while (mask) {
                                 const int i = __ffs(mask) - 1;
                                 mask &= mask - 1;
@@ -1338,6 +1344,7 @@ void tc_plan(int repr, int64_t n, int d, int k, const void *x, const void *scree
         b.cand = cv.take<int32_t>((size_t)n * (TCAND + 1));
         b.resc_rows = cv.take<int32_t>(n);
         b.fall_rows = cv.take<int32_t>(n);
+        b.fall_keys = cv.take<unsigned long long>(n);
     }
 }
 
@@ -1384,7 +1391,7 @@ int tc_assign_float(const skm_data *x, const float *C, int k, int32_t *assign, f
         rescore_kernel<uint16_t><<<gw, 256, 0, st>>>(X, d, C, b.resc_rows, b.counters, b.cand, assign);
         SKM_CUDA_TRY(launched());
         SKM_CUDA_TRY(launch_assign_exact_rows(X, 1, b.fall_rows, b.counters + 1, n, d, C, k, assign,
-                                              nullptr, st));
+                                              nullptr, b.fall_keys, st));
         if (dist) {
             assigned_dist_kernel<uint16_t><<<gw, 256, 0, st>>>(X, n, d, C, assign, dist);
             SKM_CUDA_TRY(launched());
@@ -1394,7 +1401,7 @@ int tc_assign_float(const skm_data *x, const float *C, int k, int32_t *assign, f
         rescore_kernel<float><<<gw, 256, 0, st>>>(X, d, C, b.resc_rows, b.counters, b.cand, assign);
         SKM_CUDA_TRY(launched());
         SKM_CUDA_TRY(launch_assign_exact_rows(X, 0, b.fall_rows, b.counters + 1, n, d, C, k, assign,
-                                              nullptr, st));
+                                              nullptr, b.fall_keys, st));
         if (dist) {
             assigned_dist_kernel<float><<<gw, 256, 0, st>>>(X, n, d, C, assign, dist);
             SKM_CUDA_TRY(launched());

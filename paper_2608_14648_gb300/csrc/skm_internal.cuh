@@ -111,10 +111,11 @@ cudaError_t launch_assign_exact_f32(const float *X, int64_t n, int d, const floa
                                     int32_t *assign, float *dist, cudaStream_t st);
 cudaError_t launch_assign_exact_bf16(const uint16_t *X, int64_t n, int d, const float *C, int k,
                                      int32_t *assign, float *dist, cudaStream_t st);
+// keys (optional, max_rows entries): split the centroids across the grid
 cudaError_t launch_assign_exact_rows(const void *X, int x_is_bf16, const int32_t *rows,
                                      const int32_t *count_dev, int64_t max_rows, int d,
                                      const float *C, int k, int32_t *assign, float *dist,
-                                     cudaStream_t st);
+                                     unsigned long long *keys, cudaStream_t st);
 cudaError_t launch_prune_assign(const void *X, int x_is_bf16, int64_t n, int d, const float *C,
                                 int k, const int32_t *prev, int32_t *assign, float *dist,
                                 unsigned long long *counters, cudaStream_t st);

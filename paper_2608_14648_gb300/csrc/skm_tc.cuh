@@ -27,6 +27,7 @@ struct TcAssignBufs {
     int32_t *cand = nullptr;      // F32/BF16: [n][5] screen candidates + count
     int32_t *resc_rows = nullptr;
     int32_t *fall_rows = nullptr;
+    unsigned long long *fall_keys = nullptr;  // F32/BF16: per fallback row, (dist bits, index)
 };
 
 size_t tc_screen_bytes(int repr, int64_t n, int d, const void *x);

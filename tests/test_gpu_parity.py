@@ -98,6 +98,33 @@ def test_update_f32_vs_oracle(skm):
     np.testing.assert_array_equal(C.cpu().numpy()[k - 1], C0.numpy()[k - 1])  # empty cluster kept
 
 
+@pytest.mark.parametrize("n,d,k", [(3000, 64, 300), (257, 256, 4000)])
+def test_assign_f32_screen_overflow_fallback(skm, n, d, k):
+    """Clusters of near-identical centroids (10 copies of each base point,
+    relative perturbations ~1e-6, far inside the screen's bound) leave more
+    than 4 candidates per row, so every row takes the exact fp32 fallback
+    scan, with the centroids split across the grid when the row list is short."""
+    X = _points(n, d, seed=7)
+    g = torch.Generator().manual_seed(8)
+    base = X[torch.randperm(n, generator=g)[: k // 10]]
+    C = base.repeat_interleave(10, dim=0)
+    C = (C * (1.0 + 1e-6 * torch.randn(C.shape, generator=g))).contiguous()
+    pts = skm.Points(skm.REPR_F32, X.to(DEV), d)
+    a, dist = skm.skm_assign(pts, C.to(DEV))
+    if k <= n:  # skm_fit requires k <= n; it reports how many rows fell back
+        _, _, _, _, st = skm.skm_fit(pts, k, 0, C_init=C.to(DEV), want_objective=False, want_dist=False)
+        assert st["fallback_rows"] >= n // 2
+    a_or, best, second = oracle.assign_f32(X.numpy(), C.numpy())
+    # the copies are near ties by construction, so agreement is not the test:
+    # every disagreement must sit at an oracle top-2 gap <= 1e-5, and the
+    # reported distance must be the fp32 distance to the chosen centroid
+    ag = a.cpu().numpy()
+    gap = (second - best) / np.maximum(best, 1e-30)
+    assert np.all(gap[ag != a_or] <= GAP_TOL)
+    dch = ((X.numpy().astype(np.float64) - C.numpy().astype(np.float64)[ag]) ** 2).sum(1)
+    np.testing.assert_allclose(dist.cpu().numpy(), dch, rtol=2e-5, atol=1e-6)
+
+
 def _skewed_assign(n, k, seed):
     """60% of the points in cluster 0, the rest spread over 1..k-2 (k-1 stays
     empty), and every 997th point outside [0, k) (skipped by the update)."""
