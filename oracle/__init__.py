@@ -81,6 +81,8 @@ def lib():
                 "or_mean_cov": ([vp, i64, i32, vp, vp], None),
                 "or_round_bf16": ([vp, i64, vp], None),
                 "or_sumsq_blocked": ([vp, i32], f64),
+                "or_split_empty_f32": ([vp, vp, i32, i32], i32),
+                "or_split_empty_sq8": ([vp, vp, i32, i32], i32),
             }
             for name, (args, res) in sig.items():
                 fn = getattr(L, name)
@@ -352,13 +354,30 @@ def pca_fit(X, d_out):
 # Lloyd loop (Section 2.3): iters x (STEP 2, STEP 3), then STEP 2 once more.
 # objective[t] is the objective of the assignment made at step t.
 # --------------------------------------------------------------------------
-def lloyd_f32(X, C0, iters):
+def split_empty(C, counts):
+    """Empty clusters take half of the current largest one (the library's
+    reading of splitting large clusters, Section 2.3 STEP 3); returns the new
+    centroids and the number of splits.  fp32 centroids or SQ8 codes."""
+    C = np.array(C, copy=True, order="C")
+    k, d = C.shape
+    counts = _c(counts, np.int64)
+    if C.dtype == np.uint8:
+        ns = lib().or_split_empty_sq8(_p(C), _p(counts), k, d)
+    else:
+        C = C.astype(np.float32)
+        ns = lib().or_split_empty_f32(_p(C), _p(counts), k, d)
+    return C, int(ns)
+
+
+def lloyd_f32(X, C0, iters, split=False):
     C = np.array(C0, np.float32, copy=True)
     objs = []
     for _ in range(iters):
         a, best, _ = assign_f32(X, C)
         objs.append(float(best.sum()))
         C, counts = update_f32(X, a, C)
+        if split:
+            C, _ = split_empty(C, counts)
     a, best, second = assign_f32(X, C)
     objs.append(float(best.sum()))
     return C, a, objs
@@ -376,16 +395,18 @@ def lloyd_bf16(Xb, C0, iters):
     return C, a, objs
 
 
-def lloyd_sq8(Xc, C0c, iters):
+def lloyd_sq8(Xc, C0c, iters, split=False):
     Cc = np.array(C0c, np.uint8, copy=True)
     for _ in range(iters):
         a, _ = assign_sq8(Xc, Cc)
         Cc, counts = update_sq8(Xc, a, Cc)
+        if split:
+            Cc, _ = split_empty(Cc, counts)
     a, best = assign_sq8(Xc, Cc)
     return Cc, a
 
 
-def lloyd_rbq1(codes, nx2, F, popx, d, m, C0, iters, e=None):
+def lloyd_rbq1(codes, nx2, F, popx, d, m, C0, iters, e=None, split=False):
     if e is None:
         e = rbq1_exponent(F)
     C = np.array(C0, np.float32, copy=True)
@@ -393,6 +414,8 @@ def lloyd_rbq1(codes, nx2, F, popx, d, m, C0, iters, e=None):
         prep = rbq1_centroid_sq4(C, m)
         a, _ = rbq1_assign(codes, nx2, F, popx, d, prep)
         C, counts = rbq1_update(codes, F, d, m, e, a, C)
+        if split:
+            C, _ = split_empty(C, counts)
     prep = rbq1_centroid_sq4(C, m)
     a, est = rbq1_assign(codes, nx2, F, popx, d, prep)
     return C, a

@@ -543,3 +543,67 @@ void or_round_bf16(const double *y, int64_t n, uint16_t *out) {
         out[p] = (uint16_t)(u >> 16);
     }
 }
+
+/* ------------------------------------------------------------------------ */
+/* Section 2.3 STEP 3: empty clusters are handled by splitting large ones.   */
+/* The paper only says that splitting large clusters helps; the library's   */
+/* reading: clusters left empty by an update are visited in increasing      */
+/* index order; each takes the current largest cluster L (most members,     */
+/* ties to the lowest index; nothing is done once L has fewer than 2) and   */
+/* the two become L's centroid moved symmetrically by a relative step       */
+/* eps = 2^-10 with alternating signs per dimension:                         */
+/*   new_j[i] = c_L[i] (1 + s_i eps),  new_L[i] = c_L[i] (1 - s_i eps),       */
+/*   s_i = +1 for even i, -1 for odd i  (fp32 centroids, one rounding each); */
+/* SQ8 code centroids move by one code step instead (clipped to [0, 255]).  */
+/* L keeps ceil(n_L / 2) members and j receives floor(n_L / 2) for the       */
+/* choice of later splits; the reported counts are not changed.             */
+/* ------------------------------------------------------------------------ */
+int or_split_empty_f32(float *C, const int64_t *counts, int k, int d) {
+    int64_t *w = (int64_t *)malloc(sizeof(int64_t) * (size_t)k);
+    int nsplit = 0;
+    for (int j = 0; j < k; ++j) w[j] = counts[j];
+    const float up = 1.0f + 0x1p-10f, dn = 1.0f - 0x1p-10f;
+    for (int j = 0; j < k; ++j) {
+        if (counts[j] != 0) continue;
+        int L = 0;
+        for (int t = 1; t < k; ++t)
+            if (w[t] > w[L]) L = t;
+        if (w[L] < 2) break;
+        for (int i = 0; i < d; ++i) {
+            const float c = C[(int64_t)L * d + i];
+            const int even = (i % 2) == 0;
+            C[(int64_t)j * d + i] = c * (even ? up : dn);
+            C[(int64_t)L * d + i] = c * (even ? dn : up);
+        }
+        w[j] = w[L] / 2;
+        w[L] = w[L] - w[j];
+        nsplit += 1;
+    }
+    free(w);
+    return nsplit;
+}
+
+int or_split_empty_sq8(uint8_t *C, const int64_t *counts, int k, int d) {
+    int64_t *w = (int64_t *)malloc(sizeof(int64_t) * (size_t)k);
+    int nsplit = 0;
+    for (int j = 0; j < k; ++j) w[j] = counts[j];
+    for (int j = 0; j < k; ++j) {
+        if (counts[j] != 0) continue;
+        int L = 0;
+        for (int t = 1; t < k; ++t)
+            if (w[t] > w[L]) L = t;
+        if (w[L] < 2) break;
+        for (int i = 0; i < d; ++i) {
+            const int c = C[(int64_t)L * d + i];
+            const int s = (i % 2) == 0 ? 1 : -1;
+            int a = c + s, b = c - s;
+            C[(int64_t)j * d + i] = (uint8_t)(a < 0 ? 0 : (a > 255 ? 255 : a));
+            C[(int64_t)L * d + i] = (uint8_t)(b < 0 ? 0 : (b > 255 ? 255 : b));
+        }
+        w[j] = w[L] / 2;
+        w[L] = w[L] - w[j];
+        nsplit += 1;
+    }
+    free(w);
+    return nsplit;
+}

@@ -342,3 +342,64 @@ def test_round_bf16_matches_torch_and_ties_to_even():
     # exact halfway cases: 1 + 2^-8 lies between 1 and 1 + 2^-7 -> even (1.0)
     got = oracle.round_bf16(np.array([1 + 2.0 ** -8, 1 + 3 * 2.0 ** -8, 1 + 2.0 ** -8 + 2.0 ** -30]))
     np.testing.assert_array_equal(oracle.bf16_to_f32(got), np.array([1.0, 1 + 2.0 ** -6, 1 + 2.0 ** -7], np.float32))
+
+
+# ----------------------------------------------------- empty-cluster split
+def test_split_empty_takes_the_largest_cluster_and_halves_it():
+    """Empty clusters 1 and 3 (visited in that order) each split the cluster
+    with the most members left (ties to the lowest index): 1 takes half of
+    cluster 0 (5 members: 3 stay, 2 move to 1); then cluster 0 (3) is still
+    larger than clusters 1 and 2 (2 each), so 3 splits 0 again."""
+    rng = np.random.default_rng(3)
+    C = rng.normal(size=(5, 6)).astype(np.float32)
+    counts = np.array([5, 0, 2, 0, 1], np.int64)
+    Cn, ns = oracle.split_empty(C, counts)
+    assert ns == 2
+    # untouched clusters keep their centroids
+    np.testing.assert_array_equal(Cn[2], C[2])
+    np.testing.assert_array_equal(Cn[4], C[4])
+    # the pair (1, 0) after the first split straddles the old centroid 0:
+    # each coordinate moved by a relative 2^-10 in opposite directions
+    eps = 2.0 ** -10
+    c0 = C[0].astype(np.float64)
+    first_j = c0 * np.where(np.arange(6) % 2 == 0, 1 + eps, 1 - eps)
+    np.testing.assert_allclose(Cn[1], first_j, rtol=2 ** -23)
+    # cluster 3 split the (already moved) cluster 0: midpoint of 3 and 0 is
+    # the moved centroid, and 3 differs from 1
+    moved0 = c0 * np.where(np.arange(6) % 2 == 0, 1 - eps, 1 + eps)
+    mid = (Cn[3].astype(np.float64) + Cn[0].astype(np.float64)) / 2
+    np.testing.assert_allclose(mid, moved0, rtol=1e-6)
+    assert not np.array_equal(Cn[3], Cn[1])
+
+
+def test_split_empty_tie_goes_to_lowest_index_and_singletons_are_not_split():
+    C = np.arange(12, dtype=np.float32).reshape(4, 3) + 1.0
+    Cn, ns = oracle.split_empty(C, np.array([3, 0, 3, 1], np.int64))
+    assert ns == 1
+    np.testing.assert_array_equal(Cn[2], C[2])  # tie 3 vs 3: cluster 0 is split
+    assert not np.array_equal(Cn[0], C[0])
+    Cn2, ns2 = oracle.split_empty(C, np.array([1, 0, 1, 0], np.int64))
+    assert ns2 == 0
+    np.testing.assert_array_equal(Cn2, C)
+
+
+def test_split_empty_sq8_moves_codes_by_one_step_with_clipping():
+    Cc = np.array([[0, 255, 7, 7], [9, 9, 9, 9]], np.uint8)
+    Cn, ns = oracle.split_empty(Cc, np.array([4, 0], np.int64))
+    assert ns == 1
+    np.testing.assert_array_equal(Cn[1], [1, 254, 8, 6])
+    np.testing.assert_array_equal(Cn[0], [0, 255, 6, 8])
+
+
+def test_lloyd_with_split_leaves_no_empty_cluster_on_separated_data():
+    """Two far-apart blobs and 4 centroids started inside one blob: without
+    splitting, centroids that lose every member stay empty; with splitting
+    every centroid ends with members."""
+    rng = np.random.default_rng(5)
+    X = np.concatenate([rng.normal(0, 0.1, (200, 4)), rng.normal(10, 0.1, (200, 4))]).astype(np.float32)
+    C0 = np.concatenate([X[:1] + 100, X[:1] + 101, X[200:203]]).astype(np.float32)
+    C, a, _ = oracle.lloyd_f32(X, C0, 6, split=True)
+    counts = np.bincount(a, minlength=5)
+    assert np.all(counts > 0)
+    C2, a2, _ = oracle.lloyd_f32(X, C0, 6, split=False)
+    assert np.any(np.bincount(a2, minlength=5) == 0)
