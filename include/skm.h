@@ -292,13 +292,33 @@ int skm_update_finalize(const skm_data *x, const void *partial, const int64_t *c
 typedef struct skm_fit_config {
     int32_t k;
     int32_t iters;
-    int32_t reserved[6];
+    int32_t empty_policy;  /* SKM_EMPTY_KEEP (0) or SKM_EMPTY_SPLIT (1), below */
+    int32_t reserved[5];
 } skm_fit_config;
+
+/* Empty clusters after an update (Section 2.3 STEP 3: splitting large clusters
+ * helps).  SKM_EMPTY_KEEP: an empty cluster keeps its centroid.
+ * SKM_EMPTY_SPLIT: after every update of skm_fit, skm_split_empty below. */
+enum { SKM_EMPTY_KEEP = 0, SKM_EMPTY_SPLIT = 1 };
 
 int skm_fit(const skm_fit_config *cfg, const skm_data *x, const void *C_init,
             const int64_t *init_idx, void *C_out, int32_t *assign_out, float *dist_out,
             double *objective_host, skm_stats *stats_host, void *ws, size_t ws_bytes,
             void *stream);
+
+/* Split large clusters into the empty ones (the library's reading of
+ * Section 2.3 STEP 3).  Clusters with counts[j] == 0, in increasing j, each
+ * take the current largest cluster L (most members, ties to the lowest
+ * index; nothing more happens once L has fewer than 2 members): both become
+ * L's centroid moved by a relative step of 2^-10 in opposite directions,
+ * +eps on even and -eps on odd dimensions for j (the reverse for L), one
+ * rounded fp32 multiply per element (F32/BF16/RBQ1 centroids float32[k][d]);
+ * SQ8 code centroids move by one code step instead (clipped to [0, 255]).
+ * L then counts as ceil(n_L / 2) members and j as floor(n_L / 2) for later
+ * choices; `counts` (device int64[k], from skm_update) is not modified.
+ * ws: device workspace of at least 8 k + 256 bytes.  Asynchronous. */
+int skm_split_empty(const skm_data *x, void *C_inout, const int64_t *counts, int k, void *ws,
+                    size_t ws_bytes, void *stream);
 
 /* Objective helpers (reporting, Section 4 WCSS): fp64 sum over n of
  * ||x_p - c_{a_p}||^2 with x float32 [n][d] (or bf16 bits when x_is_bf16)

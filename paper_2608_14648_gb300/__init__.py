@@ -17,12 +17,14 @@ __all__ = [
     "REPR_F32", "REPR_SQ8", "REPR_RBQ1", "REPR_BF16", "SkmError", "lib", "lib_path", "Data",
     "skm_version", "skm_kernel_launches", "skm_workspace_size", "skm_project", "skm_make_rotation", "skm_pca_fit",
     "skm_quantize", "skm_rbq1_exponent", "skm_assign", "skm_update", "skm_merge_partials",
-    "skm_update_finalize", "skm_fit", "skm_objective", "skm_sq8_decode", "EXPORTED_SYMBOLS",
+    "skm_update_finalize", "skm_fit", "skm_split_empty", "skm_objective", "skm_sq8_decode", "EXPORTED_SYMBOLS",
+    "EMPTY_KEEP", "EMPTY_SPLIT",
 ]
 
 REPR_F32, REPR_SQ8, REPR_RBQ1, REPR_BF16 = 0, 1, 2, 3
 FLAG_PRUNE = 1
 DTYPE_F32, DTYPE_BF16 = 0, 1
+EMPTY_KEEP, EMPTY_SPLIT = 0, 1
 OP_ASSIGN, OP_UPDATE, OP_FIT, OP_QUANTIZE, OP_PCA = 0, 1, 2, 3, 4
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
@@ -35,7 +37,8 @@ EXPORTED_SYMBOLS = [
     "skm_screen_prep", "skm_project", "skm_make_rotation",
     "skm_pca_fit", "skm_quantize", "skm_rbq1_exponent", "skm_assign", "skm_assign_rbq1_noalloc",
     "skm_update",
-    "skm_merge_partials", "skm_update_finalize", "skm_fit", "skm_objective", "skm_sq8_decode",
+    "skm_merge_partials", "skm_update_finalize", "skm_fit", "skm_split_empty", "skm_objective",
+    "skm_sq8_decode",
 ]
 
 
@@ -71,7 +74,8 @@ class Stats(ctypes.Structure):
 
 
 class FitConfig(ctypes.Structure):
-    _fields_ = [("k", ctypes.c_int32), ("iters", ctypes.c_int32), ("reserved", ctypes.c_int32 * 6)]
+    _fields_ = [("k", ctypes.c_int32), ("iters", ctypes.c_int32), ("empty_policy", ctypes.c_int32),
+                ("reserved", ctypes.c_int32 * 5)]
 
 
 def lib_path() -> str:
@@ -104,6 +108,7 @@ def lib():
             "skm_merge_partials": ([vp, vp, i64, i32, vp], i32),
             "skm_update_finalize": ([vp, vp, vp, i32, vp, vp], i32),
             "skm_fit": ([vp, vp, vp, vp, vp, vp, vp, vp, vp, vp, sz, vp], i32),
+            "skm_split_empty": ([vp, vp, vp, i32, vp, sz, vp], i32),
             "skm_objective": ([vp, i32, i64, i32, vp, i32, vp, vp, vp, sz, vp], i32),
             "skm_sq8_decode": ([vp, i64, i32, vp, vp, vp, vp], i32),
         }
@@ -319,8 +324,16 @@ def skm_update_finalize(pts: Points, partial, counts, C_inout, stream=None):
     return C_inout
 
 
+def skm_split_empty(pts: Points, C_inout, counts, stream=None):
+    k = C_inout.shape[0]
+    ws = _ws(8 * k + 512, pts.device)
+    _check(lib().skm_split_empty(ctypes.byref(pts.ref), _ptr(C_inout), _ptr(counts), int(k), _ptr(ws), ws.numel(),
+                                 _stream(stream)))
+    return C_inout
+
+
 def skm_fit(pts: Points, k, iters, C_init=None, init_idx=None, want_objective=True, want_dist=True,
-            ws=None, stream=None):
+            ws=None, stream=None, empty_policy=EMPTY_KEEP):
     """Returns (C, assign, dist or None, objective list or None, stats dict)."""
     dev = pts.device
     if ws is None:
@@ -333,7 +346,7 @@ def skm_fit(pts: Points, k, iters, C_init=None, init_idx=None, want_objective=Tr
     dist = torch.empty(pts.n, device=dev, dtype=torch.float32) if want_dist else None
     obj = (ctypes.c_double * (iters + 1))() if want_objective else None
     st = Stats()
-    cfg = FitConfig(int(k), int(iters))
+    cfg = FitConfig(int(k), int(iters), int(empty_policy))
     _check(lib().skm_fit(ctypes.byref(cfg), ctypes.byref(pts.ref), _ptr(C_init), _ptr(init_idx), _ptr(C),
                          _ptr(assign), _ptr(dist), obj, ctypes.byref(st), _ptr(ws), ws.numel(), _stream(stream)))
     stats = {"rescored_rows": st.rescored_rows, "fallback_rows": st.fallback_rows,

@@ -616,3 +616,94 @@ cudaError_t launch_merge(void *dst, const void *src, int64_t count, int elem_typ
 }
 
 }  // namespace skm
+
+namespace skm {
+
+// ------------------------------------------------------- empty-cluster split
+// Section 2.3 STEP 3 (splitting large clusters): clusters left empty by an
+// update, in increasing index order, each take the current largest cluster L
+// (most members, ties to the lowest index; stop once L has fewer than 2) and
+// the two become L's centroid moved by a relative 2^-10 in opposite
+// directions, the sign alternating per dimension (fp32), or by one code step
+// (SQ8, clipped).  L keeps ceil(n_L/2) members for later choices.  One block.
+constexpr int SPLIT_THREADS = 1024;
+
+template <typename T>
+__global__ void __launch_bounds__(SPLIT_THREADS) split_empty_kernel(T *__restrict__ C,
+                                                                    const int64_t *__restrict__ counts,
+                                                                    int k, int d, int64_t *__restrict__ w) {
+    __shared__ int64_t sv[SPLIT_THREADS / 32];
+    __shared__ int si[SPLIT_THREADS / 32];
+    __shared__ int sL;
+    const int tid = threadIdx.x, lane = tid & 31, wid = tid >> 5;
+    for (int j = tid; j < k; j += SPLIT_THREADS) w[j] = counts[j];
+    __syncthreads();
+    for (int j = 0; j < k; ++j) {
+        if (counts[j] != 0) continue;  // the same for every thread
+        // argmax of w, ties to the lowest index
+        int64_t bv = -1;
+        int bi = 0x7fffffff;
+        for (int t = tid; t < k; t += SPLIT_THREADS)
+            if (w[t] > bv) {
+                bv = w[t];
+                bi = t;
+            }
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) {
+            const int64_t ov = __shfl_xor_sync(0xffffffffu, bv, o);
+            const int oi = __shfl_xor_sync(0xffffffffu, bi, o);
+            if (ov > bv || (ov == bv && oi < bi)) {
+                bv = ov;
+                bi = oi;
+            }
+        }
+        if (lane == 0) {
+            sv[wid] = bv;
+            si[wid] = bi;
+        }
+        __syncthreads();
+        if (tid == 0) {
+            int64_t v = sv[0];
+            int L = si[0];
+            for (int t = 1; t < SPLIT_THREADS / 32; ++t)
+                if (sv[t] > v || (sv[t] == v && si[t] < L)) {
+                    v = sv[t];
+                    L = si[t];
+                }
+            sL = v >= 2 ? L : -1;
+        }
+        __syncthreads();
+        const int L = sL;
+        if (L < 0) break;  // the same for every thread
+        for (int i = tid; i < d; i += SPLIT_THREADS) {
+            const T c = C[(int64_t)L * d + i];
+            const bool even = (i & 1) == 0;
+            if constexpr (sizeof(T) == 1) {
+                const int s = even ? 1 : -1;
+                const int a = (int)c + s, b = (int)c - s;
+                C[(int64_t)j * d + i] = (T)(a < 0 ? 0 : (a > 255 ? 255 : a));
+                C[(int64_t)L * d + i] = (T)(b < 0 ? 0 : (b > 255 ? 255 : b));
+            } else {
+                const float up = 1.0f + 0x1p-10f, dn = 1.0f - 0x1p-10f;
+                C[(int64_t)j * d + i] = __fmul_rn(c, even ? up : dn);
+                C[(int64_t)L * d + i] = __fmul_rn(c, even ? dn : up);
+            }
+        }
+        if (tid == 0) {
+            w[j] = w[L] / 2;
+            w[L] -= w[j];
+        }
+        __syncthreads();
+    }
+}
+
+cudaError_t launch_split_empty(void *C, int code_bytes, const int64_t *counts, int k, int d,
+                               int64_t *w, cudaStream_t st) {
+    if (code_bytes == 1)
+        split_empty_kernel<uint8_t><<<1, SPLIT_THREADS, 0, st>>>(static_cast<uint8_t *>(C), counts, k, d, w);
+    else
+        split_empty_kernel<float><<<1, SPLIT_THREADS, 0, st>>>(static_cast<float *>(C), counts, k, d, w);
+    return launched();
+}
+
+}  // namespace skm

@@ -119,6 +119,7 @@ struct UpdateBufs {
     float *sumf = nullptr;    // F32/BF16: cluster sums [k][d]
     int64_t *sumi = nullptr;  // RBQ1: cluster sums [k][d + 1]; SQ8: [k][d]
     int32_t *flag = nullptr;  // raised by a streamed-sum wait that gave up
+    int64_t *wsplit = nullptr;  // empty-cluster split: working member counts [k]
 };
 
 static void plan_update(const skm_data *x, int k, Carver &cv, UpdateBufs &b) {
@@ -134,6 +135,7 @@ static void plan_update(const skm_data *x, int k, Carver &cv, UpdateBufs &b) {
     if (x->repr == SKM_REPR_SQ8) b.sumi = cv.take<int64_t>((size_t)k * x->d);
     if (x->repr == SKM_REPR_F32 || x->repr == SKM_REPR_BF16) b.sumf = cv.take<float>((size_t)k * x->d);
     b.flag = cv.take<int32_t>(1);
+    b.wsplit = cv.take<int64_t>(k);
 }
 
 struct FitBufs {
@@ -543,6 +545,8 @@ int skm_fit(const skm_fit_config *cfg, const skm_data *x, const void *C_init,
     SKM_TRY(check_k(x, k, true));
     if (cfg->iters < 0 || cfg->iters > 100000)
         return set_error(SKM_ERR_INVALID_ARG, "iters = %d", cfg->iters);
+    if (cfg->empty_policy != SKM_EMPTY_KEEP && cfg->empty_policy != SKM_EMPTY_SPLIT)
+        return set_error(SKM_ERR_INVALID_ARG, "empty_policy = %d", cfg->empty_policy);
     if (!C_out || !assign_out) return set_error(SKM_ERR_INVALID_ARG, "C_out and assign_out required");
     if (!C_init && !init_idx)
         return set_error(SKM_ERR_INVALID_ARG, "one of C_init / init_idx is required");
@@ -605,6 +609,9 @@ int skm_fit(const skm_fit_config *cfg, const skm_data *x, const void *C_init,
         }
         if (it == cfg->iters) break;
         SKM_TRY(do_update(&xd, assign, k, C_out, b.counts, nullptr, e, b.u, st));
+        if (cfg->empty_policy == SKM_EMPTY_SPLIT)
+            SKM_CUDA_TRY(launch_split_empty(C_out, x->repr == SKM_REPR_SQ8 ? 1 : 4, b.counts, k, x->d,
+                                            b.u.wsplit, st));
     }
     SKM_CUDA_TRY(cudaStreamSynchronize(st));
     skm_stats local;
@@ -626,6 +633,18 @@ int skm_fit(const skm_fit_config *cfg, const skm_data *x, const void *C_init,
             for (int j = 0; j < k; ++j) stats_host->empty_clusters += cnt[j] == 0;
         }
     }
+    return SKM_OK;
+}
+
+int skm_split_empty(const skm_data *x, void *C_inout, const int64_t *counts, int k, void *ws,
+                    size_t ws_bytes, void *stream) {
+    SKM_TRY(check_data(x, false));
+    if (!C_inout || !counts || k < 1) return set_error(SKM_ERR_INVALID_ARG, "bad arguments");
+    Carver cv(ws, ws_bytes);
+    int64_t *w = cv.take<int64_t>(k);
+    SKM_TRY(need_ws(cv, ws_bytes, ws));
+    SKM_CUDA_TRY(launch_split_empty(C_inout, x->repr == SKM_REPR_SQ8 ? 1 : 4, counts, k, x->d, w,
+                                    S(stream)));
     return SKM_OK;
 }
 

@@ -154,6 +154,9 @@ cudaError_t launch_rbq1_fq(const float *F, const int32_t *perm, const int64_t *o
 bool ring_sum_float_ok(const void *X, int x_is_bf16, int d);
 bool ring_sum_rbq1_ok(const void *codes, int d);
 bool ring_sum_sq8_ok(const void *codes, int d);
+// empty clusters take half of the largest one (w: k int64 of workspace)
+cudaError_t launch_split_empty(void *C, int code_bytes, const int64_t *counts, int k, int d,
+                               int64_t *w, cudaStream_t st);
 cudaError_t launch_ring_sum_sq8(const uint8_t *codes, int64_t n, int d, const int32_t *perm,
                                 const int32_t *scl, const int64_t *offsets, int k, int64_t *S,
                                 int32_t *flag, cudaStream_t st);

