@@ -64,6 +64,8 @@ def lib():
                 "or_assign_bf16": ([vp, i64, i32, vp, i32, vp, vp, vp], None),
                 "or_sq8_fit": ([vp, i64, i32, vp, vp], None),
                 "or_sq8_encode": ([vp, i64, i32, vp, vp, vp], None),
+                "or_sq_fit": ([vp, i64, i32, i32, vp, vp], None),
+                "or_sq_encode": ([vp, i64, i32, i32, vp, vp, vp], None),
                 "or_sq8_decode": ([vp, i64, i32, vp, vp, vp], None),
                 "or_assign_sq8": ([vp, i64, i32, vp, i32, vp, vp], None),
                 "or_update_sq8": ([vp, i64, i32, vp, i32, vp, vp], None),
@@ -146,20 +148,29 @@ def round_bf16(Y) -> np.ndarray:
 # --------------------------------------------------------------------------
 # SQ8 (Section 3.1, per-dimension parameters)
 # --------------------------------------------------------------------------
-def sq8_fit(X):
+def sq8_fit(X, bits=8):
+    """Per-dimension bias and scale of B-bit scalar codes (Section 3.1 "SQ8
+    and SQ4"): 2^B - 1 levels between the min and the max."""
     X = _c(X, np.float32)
     n, d = X.shape
     b = np.empty(d, np.float32)
     s = np.empty(d, np.float32)
-    lib().or_sq8_fit(_p(X), n, d, _p(b), _p(s))
+    if bits == 8:
+        lib().or_sq8_fit(_p(X), n, d, _p(b), _p(s))
+    else:
+        lib().or_sq_fit(_p(X), n, d, (1 << bits) - 1, _p(b), _p(s))
     return b, s
 
 
-def sq8_encode(X, b, s):
+def sq8_encode(X, b, s, bits=8):
     X = _c(X, np.float32)
     n, d = X.shape
     codes = np.empty((n, d), np.uint8)
-    lib().or_sq8_encode(_p(X), n, d, _p(_c(b, np.float32)), _p(_c(s, np.float32)), _p(codes))
+    if bits == 8:
+        lib().or_sq8_encode(_p(X), n, d, _p(_c(b, np.float32)), _p(_c(s, np.float32)), _p(codes))
+    else:
+        lib().or_sq_encode(_p(X), n, d, (1 << bits) - 1, _p(_c(b, np.float32)), _p(_c(s, np.float32)),
+                           _p(codes))
     return codes
 
 

@@ -129,7 +129,9 @@ void or_assign_bf16(const uint16_t *Xb, int64_t n, int d, const float *C, int k,
 /* with max == min gets s_i = 1.                                             */
 /* ------------------------------------------------------------------------ */
 
-void or_sq8_fit(const float *X, int64_t n, int d, float *b, float *s) {
+/* Section 3.1 "SQ8 and SQ4": B-bit codes have L = 2^B - 1 levels; per
+ * dimension b = min x, s = (max x - b) / L (s = 1 when flat). */
+void or_sq_fit(const float *X, int64_t n, int d, int levels, float *b, float *s) {
     for (int i = 0; i < d; ++i) {
         float lo = INFINITY, hi = -INFINITY;
         for (int64_t p = 0; p < n; ++p) {
@@ -137,27 +139,37 @@ void or_sq8_fit(const float *X, int64_t n, int d, float *b, float *s) {
             if (v < lo) lo = v;
             if (v > hi) hi = v;
         }
-        float sc = (hi - lo) / 255.0f;
+        float sc = (hi - lo) / (float)levels;
         if (!(sc > 0.0f)) sc = 1.0f;
         b[i] = lo;
         s[i] = sc;
     }
 }
 
+void or_sq8_fit(const float *X, int64_t n, int d, float *b, float *s) {
+    or_sq_fit(X, n, d, 255, b, s);
+}
+
 /* code = clip(round((x - b) / s), 0, 255), fp32 arithmetic, rounding half to
  * even.  Pinned: grid data reproduces codes; |decode - x| <= s/2. */
-void or_sq8_encode(const float *X, int64_t n, int d, const float *b, const float *s,
-                   uint8_t *codes) {
+void or_sq_encode(const float *X, int64_t n, int d, int levels, const float *b, const float *s,
+                  uint8_t *codes) {
+    const float top = (float)levels;
 #pragma omp parallel for schedule(static)
     for (int64_t p = 0; p < n; ++p) {
         for (int i = 0; i < d; ++i) {
             float t = (X[p * (int64_t)d + i] - b[i]) / s[i];
             float q = rintf(t);
             if (!(q >= 0.0f)) q = 0.0f;
-            if (q > 255.0f) q = 255.0f;
+            if (q > top) q = top;
             codes[p * (int64_t)d + i] = (uint8_t)q;
         }
     }
+}
+
+void or_sq8_encode(const float *X, int64_t n, int d, const float *b, const float *s,
+                   uint8_t *codes) {
+    or_sq_encode(X, n, d, 255, b, s, codes);
 }
 
 /* Reconstruction x_i ~ code_i * s_i + b_i (fp32). */

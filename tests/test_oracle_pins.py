@@ -145,6 +145,31 @@ def test_sq8_roundtrip_error_bound_and_flat_dims():
     assert np.all(err <= s.astype(np.float64) / 2 * (1 + 1e-5) + 1e-7)
 
 
+def test_sq4_grid_data_reproduces_codes_and_roundtrip_bound():
+    """4-bit codes (Section 3.1 "SQ8 and SQ4"): 15 levels between min and max.
+    Data on the grid b + s * code with s a power of two reproduces its codes;
+    generic data decodes within s/2 and uses the full 0..15 range."""
+    r = _rng(16)
+    n, d = 200, 21
+    codes = r.integers(0, 16, size=(n, d)).astype(np.uint8)
+    codes[0, :] = 0
+    codes[1, :] = 15
+    s0 = (2.0 ** -r.integers(2, 7, size=d)).astype(np.float32)
+    b0 = (r.integers(-40, 40, size=d) * s0).astype(np.float32)
+    X = (codes.astype(np.float32) * s0 + b0).astype(np.float32)
+    b, s = oracle.sq8_fit(X, bits=4)
+    np.testing.assert_array_equal(b, b0)
+    np.testing.assert_array_equal(s, s0)
+    np.testing.assert_array_equal(oracle.sq8_encode(X, b, s, bits=4), codes)
+    Y = r.standard_normal((400, 9)).astype(np.float32)
+    b, s = oracle.sq8_fit(Y, bits=4)
+    np.testing.assert_allclose(s, (Y.max(0) - Y.min(0)) / np.float32(15), rtol=1e-7)
+    c = oracle.sq8_encode(Y, b, s, bits=4)
+    assert c.max() == 15 and c.min() == 0
+    err = np.abs(oracle.sq8_decode(c, b, s).astype(np.float64) - Y)
+    assert np.all(err <= s.astype(np.float64) / 2 * (1 + 1e-5) + 1e-7)
+
+
 def test_assign_and_update_sq8_exact_integers():
     r = _rng(8)
     Xc = r.integers(0, 256, size=(120, 45)).astype(np.uint8)
