@@ -161,7 +161,10 @@ int skm_pca_fit(const float *X, int64_t n, int d, int d_out, float *mean, float 
  * ------------------------------------------------------------------------ */
 typedef struct skm_quant_params {
     int32_t fit;   /* 1: fit b,s (SQ8) or m (RBQ1) from X; 0: use supplied  */
-    int32_t reserved0;
+    int32_t bits;  /* SQ8 repr: 8 (or 0) for 8-bit codes, 4 for SQ4: 15 levels,
+                      b = min, s = (max - b) / 15, one code 0..15 per byte; SQ4
+                      codes then use every SQ8 entry point unchanged (the
+                      code-domain distance and mean are the same definitions)  */
     float *b;      /* SQ8 bias  [d] (device; output when fit, else input)    */
     float *s;      /* SQ8 scale [d]                                          */
     float *m;      /* RBQ1 mean [d]                                          */

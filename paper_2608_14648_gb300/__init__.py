@@ -61,7 +61,7 @@ class Data(ctypes.Structure):
 
 class QuantParams(ctypes.Structure):
     _fields_ = [
-        ("fit", ctypes.c_int32), ("reserved0", ctypes.c_int32), ("b", ctypes.c_void_p),
+        ("fit", ctypes.c_int32), ("bits", ctypes.c_int32), ("b", ctypes.c_void_p),
         ("s", ctypes.c_void_p), ("m", ctypes.c_void_p), ("nx2", ctypes.c_void_p),
         ("F", ctypes.c_void_p), ("popx", ctypes.c_void_p),
     ]
@@ -218,8 +218,9 @@ def skm_pca_fit(X, d_out, stream=None):
     return mean, P, w
 
 
-def skm_quantize(repr_, X, fit=True, b=None, s=None, m=None, stream=None, out=None, ws=None):
-    """SQ8 -> dict(codes, b, s); RBQ1 -> dict(codes, m, nx2, F, popx).
+def skm_quantize(repr_, X, fit=True, b=None, s=None, m=None, stream=None, out=None, ws=None, bits=8):
+    """SQ8 -> dict(codes, b, s) (bits=4: SQ4 codes 0..15, one per byte);
+    RBQ1 -> dict(codes, m, nx2, F, popx).
     `out` may supply preallocated (contiguous) output tensors by those names."""
     n, d = X.shape
     dev = X.device
@@ -232,7 +233,7 @@ def skm_quantize(repr_, X, fit=True, b=None, s=None, m=None, stream=None, out=No
         s = s if s is not None else torch.empty(d, device=dev, dtype=torch.float32)
         codes = out.get("codes")
         codes = codes if codes is not None else torch.empty(n, d, device=dev, dtype=torch.uint8)
-        qp = QuantParams(int(fit), 0, b.data_ptr(), s.data_ptr(), None, None, None, None)
+        qp = QuantParams(int(fit), int(bits), b.data_ptr(), s.data_ptr(), None, None, None, None)
         _check(lib().skm_quantize(repr_, _ptr(X), n, d, ctypes.byref(qp), _ptr(codes), _ptr(ws), ws.numel(),
                                   _stream(stream)))
         return {"codes": codes, "b": b, "s": s}

@@ -35,7 +35,8 @@ cudaError_t launch_colminmax_partial(const float *X, int64_t n, int d, float *pm
 }
 
 __global__ void sq8_params_kernel(const float *__restrict__ pmin, const float *__restrict__ pmax,
-                                  int nblk, int d, float *__restrict__ b, float *__restrict__ s) {
+                                  int nblk, int d, float levels, float *__restrict__ b,
+                                  float *__restrict__ s) {
     int c = blockIdx.x * blockDim.x + threadIdx.x;
     if (c >= d) return;
     float lo = INFINITY, hi = -INFINITY;
@@ -43,29 +44,30 @@ __global__ void sq8_params_kernel(const float *__restrict__ pmin, const float *_
         lo = fminf(lo, pmin[(int64_t)i * d + c]);
         hi = fmaxf(hi, pmax[(int64_t)i * d + c]);
     }
-    float sc = __fdiv_rn(__fsub_rn(hi, lo), 255.0f);
+    float sc = __fdiv_rn(__fsub_rn(hi, lo), levels);
     if (!(sc > 0.0f)) sc = 1.0f;
     b[c] = lo;
     s[c] = sc;
 }
 
-cudaError_t launch_sq8_params(const float *pmin, const float *pmax, int nblk, int d, float *b,
-                              float *s, cudaStream_t st) {
-    sq8_params_kernel<<<(d + 127) / 128, 128, 0, st>>>(pmin, pmax, nblk, d, b, s);
+cudaError_t launch_sq8_params(const float *pmin, const float *pmax, int nblk, int d, int levels,
+                              float *b, float *s, cudaStream_t st) {
+    sq8_params_kernel<<<(d + 127) / 128, 128, 0, st>>>(pmin, pmax, nblk, d, (float)levels, b, s);
     return launched();
 }
 
-// code = clip(rint((x - b) / s), 0, 255); 16 elements per thread per step.
-__device__ __forceinline__ uint32_t sq8_code(float x, float b, float s) {
+// code = clip(rint((x - b) / s), 0, L) (L = 255 for 8-bit, 15 for 4-bit
+// codes, one code per byte); 16 elements per thread per step.
+__device__ __forceinline__ uint32_t sq8_code(float x, float b, float s, float top) {
     float q = rintf(__fdiv_rn(__fsub_rn(x, b), s));
     q = (q >= 0.0f) ? q : 0.0f;
-    q = fminf(q, 255.0f);
+    q = fminf(q, top);
     return (uint32_t)q;
 }
 
 __global__ void sq8_encode_vec_kernel(const float4 *__restrict__ X, int64_t n16, int d,
                                       const float *__restrict__ b, const float *__restrict__ s,
-                                      uint4 *__restrict__ out) {
+                                      float top, uint4 *__restrict__ out) {
     // requires d % 16 == 0: a 16-element chunk never crosses a row
     for (int64_t t = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; t < n16;
          t += (int64_t)gridDim.x * blockDim.x) {
@@ -77,9 +79,9 @@ __global__ void sq8_encode_vec_kernel(const float4 *__restrict__ X, int64_t n16,
 #pragma unroll
         for (int q = 0; q < 4; ++q) {
             const int c = c0 + 4 * q;
-            w[q] = sq8_code(v[q].x, b[c], s[c]) | (sq8_code(v[q].y, b[c + 1], s[c + 1]) << 8) |
-                   (sq8_code(v[q].z, b[c + 2], s[c + 2]) << 16) |
-                   (sq8_code(v[q].w, b[c + 3], s[c + 3]) << 24);
+            w[q] = sq8_code(v[q].x, b[c], s[c], top) | (sq8_code(v[q].y, b[c + 1], s[c + 1], top) << 8) |
+                   (sq8_code(v[q].z, b[c + 2], s[c + 2], top) << 16) |
+                   (sq8_code(v[q].w, b[c + 3], s[c + 3], top) << 24);
         }
         out[t] = make_uint4(w[0], w[1], w[2], w[3]);
     }
@@ -87,11 +89,11 @@ __global__ void sq8_encode_vec_kernel(const float4 *__restrict__ X, int64_t n16,
 
 __global__ void sq8_encode_scalar_kernel(const float *__restrict__ X, int64_t total, int d,
                                          const float *__restrict__ b, const float *__restrict__ s,
-                                         uint8_t *__restrict__ out) {
+                                         float top, uint8_t *__restrict__ out) {
     for (int64_t t = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; t < total;
          t += (int64_t)gridDim.x * blockDim.x) {
         const int c = (int)(t % d);
-        out[t] = (uint8_t)sq8_code(X[t], b[c], s[c]);
+        out[t] = (uint8_t)sq8_code(X[t], b[c], s[c], top);
     }
 }
 
@@ -104,14 +106,15 @@ static int grid_for(int64_t work, int threads) {
 }
 
 cudaError_t launch_sq8_encode(const float *X, int64_t n, int d, const float *b, const float *s,
-                              uint8_t *codes, cudaStream_t st) {
+                              int levels, uint8_t *codes, cudaStream_t st) {
     const int64_t total = n * d;
+    const float top = (float)levels;
     if (d % 16 == 0 && (((uintptr_t)X | (uintptr_t)codes) & 15) == 0) {
         const int64_t n16 = total / 16;
         sq8_encode_vec_kernel<<<grid_for(n16, 256), 256, 0, st>>>(
-            reinterpret_cast<const float4 *>(X), n16, d, b, s, reinterpret_cast<uint4 *>(codes));
+            reinterpret_cast<const float4 *>(X), n16, d, b, s, top, reinterpret_cast<uint4 *>(codes));
     } else {
-        sq8_encode_scalar_kernel<<<grid_for(total, 256), 256, 0, st>>>(X, total, d, b, s, codes);
+        sq8_encode_scalar_kernel<<<grid_for(total, 256), 256, 0, st>>>(X, total, d, b, s, top, codes);
     }
     return launched();
 }

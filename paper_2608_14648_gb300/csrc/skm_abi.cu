@@ -423,12 +423,15 @@ int skm_quantize(int repr, const float *X, int64_t n, int d, skm_quant_params *q
     const int nblk = (int)std::min<int64_t>(RED_BLOCKS, n);
     if (repr == SKM_REPR_SQ8) {
         if (!qp->b || !qp->s) return set_error(SKM_ERR_INVALID_ARG, "SQ8 needs b and s");
+        if (qp->bits != 0 && qp->bits != 8 && qp->bits != 4)
+            return set_error(SKM_ERR_INVALID_ARG, "bits = %d (0, 4 or 8)", qp->bits);
+        const int levels = qp->bits == 4 ? 15 : 255;
         if (qp->fit) {
             SKM_TRY(need_ws(cv, ws_bytes, ws));
             SKM_CUDA_TRY(launch_colminmax_partial(X, n, d, pmin, pmax, nblk, st));
-            SKM_CUDA_TRY(launch_sq8_params(pmin, pmax, nblk, d, qp->b, qp->s, st));
+            SKM_CUDA_TRY(launch_sq8_params(pmin, pmax, nblk, d, levels, qp->b, qp->s, st));
         }
-        SKM_CUDA_TRY(launch_sq8_encode(X, n, d, qp->b, qp->s, static_cast<uint8_t *>(codes), st));
+        SKM_CUDA_TRY(launch_sq8_encode(X, n, d, qp->b, qp->s, levels, static_cast<uint8_t *>(codes), st));
         return SKM_OK;
     }
     if (repr == SKM_REPR_RBQ1) {

@@ -83,10 +83,11 @@ struct Rbq1CInfo {
 // quantize / encode
 cudaError_t launch_colminmax_partial(const float *X, int64_t n, int d, float *pmin, float *pmax,
                                      int nblk, cudaStream_t st);
-cudaError_t launch_sq8_params(const float *pmin, const float *pmax, int nblk, int d, float *b,
-                              float *s, cudaStream_t st);
+// levels L = 2^bits - 1 (255 for SQ8, 15 for SQ4)
+cudaError_t launch_sq8_params(const float *pmin, const float *pmax, int nblk, int d, int levels,
+                              float *b, float *s, cudaStream_t st);
 cudaError_t launch_sq8_encode(const float *X, int64_t n, int d, const float *b, const float *s,
-                              uint8_t *codes, cudaStream_t st);
+                              int levels, uint8_t *codes, cudaStream_t st);
 cudaError_t launch_sq8_decode(const uint8_t *codes, int64_t n, int d, const float *b,
                               const float *s, float *Y, cudaStream_t st);
 cudaError_t launch_colsum_partial(const float *X, int64_t n, int d, double *psum, int nblk,

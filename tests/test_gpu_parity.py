@@ -523,3 +523,25 @@ def test_fit_f32_with_split_vs_oracle(skm):
     _, a0, _, _, _ = skm.skm_fit(pts, k, iters, init_idx=idx.to(DEV))
     empty = lambda v: int((np.bincount(v, minlength=k) == 0).sum())  # noqa: E731
     assert empty(a.cpu().numpy()) < empty(a0.cpu().numpy())
+
+
+# ------------------------------------------------------------------- SQ4
+@pytest.mark.parametrize("n,d,k", [(3000, 64, 40), (1500, 1024, 33), (777, 33, 7)])
+def test_sq4_quantize_assign_update_fit_bitexact(skm, n, d, k):
+    """4-bit codes through the SQ8 entry points: encode, exact code-domain
+    assignment and update, and a whole Lloyd trajectory, against the oracle."""
+    X = _points(n, d, seed=n + 4)
+    q = skm.skm_quantize(skm.REPR_SQ8, X.to(DEV), bits=4)
+    b, s = oracle.sq8_fit(X.numpy(), bits=4)
+    np.testing.assert_array_equal(q["b"].cpu().numpy(), b)
+    np.testing.assert_array_equal(q["s"].cpu().numpy(), s)
+    codes = q["codes"].cpu().numpy()
+    np.testing.assert_array_equal(codes, oracle.sq8_encode(X.numpy(), b, s, bits=4))
+    assert codes.max() <= 15
+    pts = skm.Points(skm.REPR_SQ8, q["codes"], d)
+    idx = synth.forgy_indices(n, k, seed=4)
+    C, a, dist, _, _ = skm.skm_fit(pts, k, 4, init_idx=idx.to(DEV))
+    Co, ao = oracle.lloyd_sq8(codes, codes[idx.numpy()], 4)
+    np.testing.assert_array_equal(a.cpu().numpy(), ao)
+    np.testing.assert_array_equal(C.cpu().numpy(), Co)
+    assert C.cpu().numpy().max() <= 15
