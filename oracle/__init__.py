@@ -84,6 +84,7 @@ def lib():
                 "or_round_bf16": ([vp, i64, vp], None),
                 "or_sumsq_blocked": ([vp, i32], f64),
                 "or_split_empty_f32": ([vp, vp, i32, i32], i32),
+                "or_hadamard_rotate": ([vp, i64, i32, vp, vp, i32, vp], None),
                 "or_split_empty_sq8": ([vp, vp, i32, i32], i32),
             }
             for name, (args, res) in sig.items():
@@ -365,6 +366,20 @@ def pca_fit(X, d_out):
 # Lloyd loop (Section 2.3): iters x (STEP 2, STEP 3), then STEP 2 once more.
 # objective[t] is the objective of the assignment made at step t.
 # --------------------------------------------------------------------------
+def hadamard_rotate(X, sigma, mean=None):
+    """y = H_D diag(sigma) [x - mean; 0] / sqrt(D), D = len(sigma) (a power of
+    two >= d), in fp64 (fast Walsh-Hadamard transform), rounded to fp32."""
+    X = _c(X, np.float32)
+    n, d = X.shape
+    sigma = _c(sigma, np.float32)
+    D = sigma.shape[0]
+    assert D >= d and D & (D - 1) == 0
+    Y = np.empty((n, D), np.float32)
+    lib().or_hadamard_rotate(_p(X), n, d, _p(_c(mean, np.float32)) if mean is not None else None, _p(sigma), D,
+                             _p(Y))
+    return Y
+
+
 def split_empty(C, counts):
     """Empty clusters take half of the current largest one (the library's
     reading of splitting large clusters, Section 2.3 STEP 3); returns the new

@@ -619,3 +619,35 @@ int or_split_empty_sq8(uint8_t *C, const int64_t *counts, int k, int d) {
     free(w);
     return nsplit;
 }
+
+/* ------------------------------------------------------------------------ */
+/* Randomized Hadamard rotation (a structured random orthogonal transform,   */
+/* used in place of a dense random rotation before RabitQ / SuperKMeans,    */
+/* Section 3.1): y = (1/sqrt(D)) H_D diag(sigma) [x - mean ; 0], with D the  */
+/* smallest power of two >= d (the row is zero-padded), H_D the Sylvester    */
+/* Hadamard matrix (H_1 = 1, H_2m = [[H_m, H_m], [H_m, -H_m]]) and sigma a   */
+/* given +-1 vector.  fp64 in-place fast Walsh-Hadamard transform, then one */
+/* rounding to fp32.                                                         */
+/* ------------------------------------------------------------------------ */
+void or_hadamard_rotate(const float *X, int64_t n, int d, const float *mean, const float *sigma,
+                        int D, float *Y) {
+    const double scale = 1.0 / sqrt((double)D);
+#pragma omp parallel for schedule(static)
+    for (int64_t p = 0; p < n; ++p) {
+        double *v = (double *)malloc(sizeof(double) * (size_t)D);
+        for (int i = 0; i < D; ++i) {
+            double x = 0.0;
+            if (i < d) x = (double)X[p * (int64_t)d + i] - (mean ? (double)mean[i] : 0.0);
+            v[i] = x * (double)sigma[i];
+        }
+        for (int h = 1; h < D; h <<= 1)
+            for (int i = 0; i < D; i += 2 * h)
+                for (int j = i; j < i + h; ++j) {
+                    const double a = v[j], b = v[j + h];
+                    v[j] = a + b;
+                    v[j + h] = a - b;
+                }
+        for (int i = 0; i < D; ++i) Y[p * (int64_t)D + i] = (float)(v[i] * scale);
+        free(v);
+    }
+}

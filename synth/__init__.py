@@ -122,6 +122,13 @@ def gmm_points(
     return out
 
 
+def hadamard_signs(D: int, seed: int) -> torch.Tensor:
+    """Seeded +-1 vector of length D (float32, CPU) for a randomized Hadamard
+    rotation."""
+    g = _generator(seed + 3, "cpu")
+    return (torch.randint(0, 2, (D,), generator=g) * 2 - 1).to(torch.float32)
+
+
 def forgy_indices(n: int, k: int, seed: int) -> torch.Tensor:
     """First k entries of a seeded uniform permutation of range(n) (int64, CPU)."""
     g = _generator(seed + 2, "cpu")

@@ -428,3 +428,38 @@ def test_lloyd_with_split_leaves_no_empty_cluster_on_separated_data():
     assert np.all(counts > 0)
     C2, a2, _ = oracle.lloyd_f32(X, C0, 6, split=False)
     assert np.any(np.bincount(a2, minlength=5) == 0)
+
+
+# -------------------------------------------------- randomized Hadamard rotation
+def test_hadamard_rotate_small_cases_by_hand():
+    # D = 2: (x0 s0 + x1 s1, x0 s0 - x1 s1) / sqrt(2)
+    X = np.array([[3.0, 1.0]], np.float32)
+    Y = oracle.hadamard_rotate(X, np.array([1.0, -1.0], np.float32))
+    np.testing.assert_allclose(Y[0], np.array([2.0, 4.0]) / np.sqrt(2), rtol=1e-7)
+    # D = 4 with padding of a 3-dimensional row and a mean: rows of H_4 are
+    # (1,1,1,1), (1,-1,1,-1), (1,1,-1,-1), (1,-1,-1,1)
+    X = np.array([[2.0, 5.0, -1.0]], np.float32)
+    mean = np.array([1.0, 1.0, 1.0], np.float32)
+    s = np.array([1.0, 1.0, -1.0, 1.0], np.float32)
+    v = np.array([1.0, 4.0, 2.0, 0.0])  # (x - mean) * sigma, padded
+    H4 = np.array([[1, 1, 1, 1], [1, -1, 1, -1], [1, 1, -1, -1], [1, -1, -1, 1]], np.float64)
+    np.testing.assert_allclose(oracle.hadamard_rotate(X, s, mean)[0], H4 @ v / 2.0, rtol=1e-7)
+
+
+def test_hadamard_rotate_is_orthogonal_and_preserves_distances():
+    r = _rng(21)
+    X = r.standard_normal((50, 100)).astype(np.float32)
+    s = np.where(r.random(128) < 0.5, -1.0, 1.0).astype(np.float32)
+    Y = oracle.hadamard_rotate(X, s).astype(np.float64)
+    assert Y.shape == (50, 128)
+    Xd = X.astype(np.float64)
+    np.testing.assert_allclose(np.linalg.norm(Y, axis=1), np.linalg.norm(Xd, axis=1), rtol=1e-6)
+    dX = np.linalg.norm(Xd[:, None] - Xd[None], axis=2)
+    dY = np.linalg.norm(Y[:, None] - Y[None], axis=2)
+    np.testing.assert_allclose(dY, dX, rtol=1e-5, atol=1e-5)
+    # the transform of the unit vectors e_i is the i-th column of H D / sqrt(D):
+    # entries +-1/sqrt(D), columns mutually orthogonal
+    E = np.eye(128, dtype=np.float32)
+    T = oracle.hadamard_rotate(E, s).astype(np.float64)
+    np.testing.assert_allclose(np.abs(T), 1 / np.sqrt(128), rtol=1e-7)
+    np.testing.assert_allclose(T @ T.T, np.eye(128), atol=1e-6)
