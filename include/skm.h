@@ -128,6 +128,18 @@ size_t skm_workspace_size(int op, const skm_data *x, int k);
 int skm_project(const float *X, int64_t n, int d, const float *mean, const float *P,
                 int d_out, int out_dtype, void *Y, void *stream);
 
+/* Randomized Hadamard rotation (a structured random orthogonal transform in
+ * place of a dense random rotation before RabitQ / SuperKMeans, Section 3.1;
+ * O(D log D) per point): Y = (1/sqrt(D)) H_D diag(sigma) [X - mean; 0] with
+ * H_D the Sylvester Hadamard matrix (H_1 = 1, H_2m = [[H_m, H_m], [H_m, -H_m]]),
+ * every row zero-padded from d to D dimensions.  D: power of two, max(32, d)
+ * <= D <= 4096.  sigma: device float32[D] of +1/-1 (the random draw, supplied
+ * by the caller); mean: device float32[d] or NULL.  Y (device): float32 or bf16
+ * [n][D] (out_dtype, bf16 rounded to nearest even).  fp32 arithmetic.
+ * Distances are preserved up to rounding.  Asynchronous. */
+int skm_project_hadamard(const float *X, int64_t n, int d, const float *mean, const float *sigma,
+                         int D, int out_dtype, void *Y, void *stream);
+
 /* Haar-random orthogonal d x d matrix (HOST helper, host output P_host[d][d],
  * float32 row-major): Householder QR of a Gaussian matrix drawn with
  * Philox4x32-10 + Box-Muller from `seed`, signs fixed so R has a positive

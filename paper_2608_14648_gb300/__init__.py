@@ -15,7 +15,8 @@ import torch
 
 __all__ = [
     "REPR_F32", "REPR_SQ8", "REPR_RBQ1", "REPR_BF16", "SkmError", "lib", "lib_path", "Data",
-    "skm_version", "skm_kernel_launches", "skm_workspace_size", "skm_project", "skm_make_rotation", "skm_pca_fit",
+    "skm_version", "skm_kernel_launches", "skm_workspace_size", "skm_project", "skm_project_hadamard",
+    "skm_make_rotation", "skm_pca_fit",
     "skm_quantize", "skm_rbq1_exponent", "skm_assign", "skm_update", "skm_merge_partials",
     "skm_update_finalize", "skm_fit", "skm_split_empty", "skm_objective", "skm_sq8_decode", "EXPORTED_SYMBOLS",
     "EMPTY_KEEP", "EMPTY_SPLIT",
@@ -34,7 +35,7 @@ _lib = None
 # Every entry point declared in include/skm.h.
 EXPORTED_SYMBOLS = [
     "skm_last_error", "skm_version", "skm_kernel_launches", "skm_workspace_size", "skm_screen_bytes",
-    "skm_screen_prep", "skm_project", "skm_make_rotation",
+    "skm_screen_prep", "skm_project", "skm_project_hadamard", "skm_make_rotation",
     "skm_pca_fit", "skm_quantize", "skm_rbq1_exponent", "skm_assign", "skm_assign_rbq1_noalloc",
     "skm_update",
     "skm_merge_partials", "skm_update_finalize", "skm_fit", "skm_split_empty", "skm_objective",
@@ -99,6 +100,7 @@ def lib():
             "skm_screen_prep": ([vp, vp, sz, vp], i32),
             "skm_project": ([vp, i64, i32, vp, vp, i32, i32, vp, vp], i32),
             "skm_make_rotation": ([u64, i32, vp], i32),
+            "skm_project_hadamard": ([vp, i64, i32, vp, vp, i32, i32, vp, vp], i32),
             "skm_pca_fit": ([vp, i64, i32, i32, vp, vp, vp, vp, sz, vp], i32),
             "skm_quantize": ([i32, vp, i64, i32, vp, vp, vp, sz, vp], i32),
             "skm_rbq1_exponent": ([vp, i64, vp, vp, sz, vp], i32),
@@ -197,6 +199,16 @@ def skm_project(X, P, mean=None, out_dtype=DTYPE_F32, stream=None):
     d_out = P.shape[1]
     Y = torch.empty(n, d_out, device=X.device, dtype=torch.float32 if out_dtype == DTYPE_F32 else torch.bfloat16)
     _check(lib().skm_project(_ptr(X), n, d, _ptr(mean), _ptr(P), d_out, out_dtype, _ptr(Y), _stream(stream)))
+    return Y
+
+
+def skm_project_hadamard(X, sigma, mean=None, out_dtype=DTYPE_F32, stream=None):
+    """Randomized Hadamard rotation; sigma: device float32 [D] of +-1 (D a power of two >= d)."""
+    n, d = X.shape
+    D = sigma.numel()
+    Y = torch.empty(n, D, device=X.device, dtype=torch.float32 if out_dtype == DTYPE_F32 else torch.bfloat16)
+    _check(lib().skm_project_hadamard(_ptr(X), n, d, _ptr(mean), _ptr(sigma), int(D), out_dtype, _ptr(Y),
+                                      _stream(stream)))
     return Y
 
 

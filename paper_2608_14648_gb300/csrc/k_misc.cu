@@ -321,3 +321,125 @@ cudaError_t launch_cov_reduce(const double *partial, int splits, int d, double *
 }
 
 }  // namespace skm
+
+namespace skm {
+
+// -------------------------------------------------- randomized Hadamard rotation
+// y = (1/sqrt(D)) H_D diag(sigma) [x - mean; 0] (a structured random
+// orthogonal transform, Section 3.1's rotation before RabitQ / SuperKMeans,
+// O(D log D) per row instead of a D x D product).  Element i of the padded
+// row lives in lane i % 32, register i / 32 of one warp; the Walsh-Hadamard
+// butterflies over the register bits run inside each lane and those over the
+// lane bits through __shfl_xor_sync.  The transform is a product of
+// independent per-bit butterflies, so their order does not change the
+// result beyond rounding.  D <= 1024 here; 2048 and 4096 use shared memory.
+template <int J>
+__global__ void __launch_bounds__(256) hadamard_warp_kernel(const float *__restrict__ X, int64_t n, int d,
+                                                            const float *__restrict__ mean,
+                                                            const float *__restrict__ sigma, float scale,
+                                                            int out_bf16, void *__restrict__ Y) {
+    constexpr int D = 32 * J;
+    const int lane = threadIdx.x & 31;
+    const int64_t warp = (blockIdx.x * (int64_t)blockDim.x + threadIdx.x) >> 5;
+    const int64_t nw = ((int64_t)gridDim.x * blockDim.x) >> 5;
+    float sg[J], mu[J];
+#pragma unroll
+    for (int j = 0; j < J; ++j) {
+        const int i = lane + 32 * j;
+        sg[j] = __ldg(sigma + i);
+        mu[j] = (mean && i < d) ? __ldg(mean + i) : 0.0f;
+    }
+    for (int64_t r = warp; r < n; r += nw) {
+        float v[J];
+#pragma unroll
+        for (int j = 0; j < J; ++j) {
+            const int i = lane + 32 * j;
+            const float x = i < d ? __ldg(X + r * d + i) : 0.0f;
+            v[j] = __fmul_rn(__fsub_rn(x, mu[j]), sg[j]);
+        }
+#pragma unroll
+        for (int h = 1; h < J; h <<= 1)
+#pragma unroll
+            for (int j = 0; j < J; ++j)
+                if ((j & h) == 0) {
+                    const float a = v[j], b = v[j + h];
+                    v[j] = __fadd_rn(a, b);
+                    v[j + h] = __fsub_rn(a, b);
+                }
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1)
+#pragma unroll
+            for (int j = 0; j < J; ++j) {
+                const float p = __shfl_xor_sync(0xffffffffu, v[j], o);
+                v[j] = (lane & o) ? __fsub_rn(p, v[j]) : __fadd_rn(v[j], p);
+            }
+#pragma unroll
+        for (int j = 0; j < J; ++j) {
+            const int i = lane + 32 * j;
+            const float y = __fmul_rn(v[j], scale);
+            if (out_bf16)
+                reinterpret_cast<__nv_bfloat16 *>(Y)[r * D + i] = __float2bfloat16_rn(y);
+            else
+                reinterpret_cast<float *>(Y)[r * D + i] = y;
+        }
+    }
+}
+
+// D = 2048 or 4096: one block per row, the row in shared memory.
+__global__ void __launch_bounds__(512) hadamard_block_kernel(const float *__restrict__ X, int64_t n, int d, int D,
+                                                             const float *__restrict__ mean,
+                                                             const float *__restrict__ sigma, float scale,
+                                                             int out_bf16, void *__restrict__ Y) {
+    __shared__ float v[4096];
+    for (int64_t r = blockIdx.x; r < n; r += gridDim.x) {
+        __syncthreads();
+        for (int i = threadIdx.x; i < D; i += blockDim.x) {
+            const float x = i < d ? __ldg(X + r * d + i) : 0.0f;
+            const float m = (mean && i < d) ? __ldg(mean + i) : 0.0f;
+            v[i] = __fmul_rn(__fsub_rn(x, m), __ldg(sigma + i));
+        }
+        for (int h = 1; h < D; h <<= 1) {
+            __syncthreads();
+            for (int t = threadIdx.x; t < D / 2; t += blockDim.x) {
+                const int j = (t / h) * 2 * h + (t % h);
+                const float a = v[j], b = v[j + h];
+                v[j] = __fadd_rn(a, b);
+                v[j + h] = __fsub_rn(a, b);
+            }
+        }
+        __syncthreads();
+        for (int i = threadIdx.x; i < D; i += blockDim.x) {
+            const float y = __fmul_rn(v[i], scale);
+            if (out_bf16)
+                reinterpret_cast<__nv_bfloat16 *>(Y)[r * D + i] = __float2bfloat16_rn(y);
+            else
+                reinterpret_cast<float *>(Y)[r * D + i] = y;
+        }
+    }
+}
+
+cudaError_t launch_hadamard(const float *X, int64_t n, int d, const float *mean, const float *sigma, int D,
+                            int out_bf16, void *Y, cudaStream_t st) {
+    if (n == 0) return cudaSuccess;
+    const float scale = (float)(1.0 / sqrt((double)D));
+    if (D <= 1024) {
+        int64_t blocks = (n * 32 + 255) / 256;
+        if (blocks > 152 * 8) blocks = 152 * 8;
+        const int g = (int)blocks;
+        switch (D) {
+        case 32: hadamard_warp_kernel<1><<<g, 256, 0, st>>>(X, n, d, mean, sigma, scale, out_bf16, Y); break;
+        case 64: hadamard_warp_kernel<2><<<g, 256, 0, st>>>(X, n, d, mean, sigma, scale, out_bf16, Y); break;
+        case 128: hadamard_warp_kernel<4><<<g, 256, 0, st>>>(X, n, d, mean, sigma, scale, out_bf16, Y); break;
+        case 256: hadamard_warp_kernel<8><<<g, 256, 0, st>>>(X, n, d, mean, sigma, scale, out_bf16, Y); break;
+        case 512: hadamard_warp_kernel<16><<<g, 256, 0, st>>>(X, n, d, mean, sigma, scale, out_bf16, Y); break;
+        case 1024: hadamard_warp_kernel<32><<<g, 256, 0, st>>>(X, n, d, mean, sigma, scale, out_bf16, Y); break;
+        default: return cudaErrorInvalidValue;
+        }
+        return launched();
+    }
+    int64_t blocks = n < 152 * 4 ? n : 152 * 4;
+    hadamard_block_kernel<<<(int)blocks, 512, 0, st>>>(X, n, d, D, mean, sigma, scale, out_bf16, Y);
+    return launched();
+}
+
+}  // namespace skm

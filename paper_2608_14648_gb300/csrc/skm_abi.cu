@@ -355,6 +355,18 @@ int skm_project(const float *X, int64_t n, int d, const float *mean, const float
     return SKM_OK;
 }
 
+int skm_project_hadamard(const float *X, int64_t n, int d, const float *mean, const float *sigma, int D,
+                         int out_dtype, void *Y, void *stream) {
+    if (!X || !sigma || !Y) return set_error(SKM_ERR_INVALID_ARG, "NULL pointer");
+    if (n < 1 || d < 1 || d > MAX_D) return set_error(SKM_ERR_INVALID_ARG, "bad shape n=%lld d=%d", (long long)n, d);
+    if (D < 32 || D > 4096 || (D & (D - 1)) != 0 || D < d)
+        return set_error(SKM_ERR_INVALID_ARG, "D = %d must be a power of two in [max(32, d), 4096]", D);
+    if (out_dtype != SKM_DTYPE_F32 && out_dtype != SKM_DTYPE_BF16)
+        return set_error(SKM_ERR_INVALID_ARG, "bad out_dtype %d", out_dtype);
+    SKM_CUDA_TRY(launch_hadamard(X, n, d, mean, sigma, D, out_dtype == SKM_DTYPE_BF16, Y, S(stream)));
+    return SKM_OK;
+}
+
 int skm_make_rotation(uint64_t seed, int d, float *P_host) {
     if (!P_host || d < 1 || d > MAX_D) return set_error(SKM_ERR_INVALID_ARG, "bad arguments");
     std::vector<double> A((size_t)d * d);

@@ -155,6 +155,9 @@ cudaError_t launch_rbq1_fq(const float *F, const int32_t *perm, const int64_t *o
 bool ring_sum_float_ok(const void *X, int x_is_bf16, int d);
 bool ring_sum_rbq1_ok(const void *codes, int d);
 bool ring_sum_sq8_ok(const void *codes, int d);
+// y = H_D diag(sigma) [x - mean; 0] / sqrt(D), D a power of two in [32, 4096]
+cudaError_t launch_hadamard(const float *X, int64_t n, int d, const float *mean, const float *sigma, int D,
+                            int out_bf16, void *Y, cudaStream_t st);
 // empty clusters take half of the largest one (w: k int64 of workspace)
 cudaError_t launch_split_empty(void *C, int code_bytes, const int64_t *counts, int k, int d,
                                int64_t *w, cudaStream_t st);

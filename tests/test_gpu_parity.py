@@ -545,3 +545,21 @@ def test_sq4_quantize_assign_update_fit_bitexact(skm, n, d, k):
     np.testing.assert_array_equal(a.cpu().numpy(), ao)
     np.testing.assert_array_equal(C.cpu().numpy(), Co)
     assert C.cpu().numpy().max() <= 15
+
+
+# ------------------------------------------------ randomized Hadamard rotation
+@pytest.mark.parametrize("n,d,D", [(1000, 33, 64), (777, 100, 128), (3000, 768, 1024), (500, 1024, 1024),
+                                   (300, 2000, 2048), (64, 4096, 4096), (50, 20, 32)])
+def test_project_hadamard_vs_oracle(skm, n, d, D):
+    X = _points(n, d, seed=d + 1)
+    sigma = synth.hadamard_signs(D, seed=d)
+    mean = X.mean(0) if d % 2 else None
+    Y = skm.skm_project_hadamard(X.to(DEV), sigma.to(DEV), None if mean is None else mean.to(DEV))
+    Yo = oracle.hadamard_rotate(X.numpy(), sigma.numpy(), None if mean is None else mean.numpy())
+    Yg = Y.cpu().numpy().astype(np.float64)
+    err = np.linalg.norm(Yg - Yo, axis=1) / np.maximum(np.linalg.norm(Yo, axis=1), 1e-30)
+    assert err.max() <= 2e-6
+    # bf16 output: the fp32 result rounded to nearest even
+    Yb = skm.skm_project_hadamard(X.to(DEV), sigma.to(DEV), None if mean is None else mean.to(DEV),
+                                  out_dtype=skm.DTYPE_BF16).float().cpu().numpy()
+    assert np.all(np.abs(Yb - Yo) <= 2.0 ** -8 * np.abs(Yo) + 1e-6)
