@@ -445,3 +445,86 @@ def lloyd_rbq1(codes, nx2, F, popx, d, m, C0, iters, e=None, split=False):
     prep = rbq1_centroid_sq4(C, m)
     a, est = rbq1_assign(codes, nx2, F, popx, d, prep)
     return C, a
+
+
+# --------------------------------------------------------------------------
+# Hierarchical k-means (the paper's MESO- and FINE-CLUSTERING, with the
+# optional refinement iteration of vanilla k-means).
+# --------------------------------------------------------------------------
+def fine_counts(sizes, k):
+    """Fine clusters per meso cluster: k apportioned proportionally to the
+    meso sizes n_i (floor of k n_i / N, the remaining clusters to the largest
+    remainders k n_i mod N, ties to the lower index); a non-empty meso cluster
+    left with none takes one from the cluster with the most (ties to the lower
+    index).  Empty meso clusters get none.  The paper states sqrt(n_i) fine
+    clusters per meso cluster; this reading keeps the total at the requested k."""
+    sizes = [int(v) for v in sizes]
+    N = sum(sizes)
+    m = len(sizes)
+    kk = [k * v // N for v in sizes]
+    rem = [k * v % N for v in sizes]
+    left = k - sum(kk)
+    order = sorted(range(m), key=lambda i: (-rem[i], i))
+    for i in order[:left]:
+        kk[i] += 1
+    for i in range(m):
+        if sizes[i] > 0 and kk[i] == 0:
+            j = min(range(m), key=lambda t: (-kk[t], t))
+            kk[j] -= 1
+            kk[i] = 1
+    return kk
+
+
+def fine_init_positions(n_i, k_i):
+    """Positions (in the meso cluster's members, increasing point index) of the
+    initial fine centroids: floor(t n_i / k_i), t < k_i."""
+    return [t * n_i // k_i for t in range(k_i)]
+
+
+def hierarchical(kind, data, k, m, meso_init, meso_iters, fine_iters, refine=False):
+    """kind 'f32' (data = X), 'sq8' (data = codes) or 'rbq1' (data = dict of
+    codes, nx2, F, popx, d, m, e).  Returns (centroids [k], assignments [n],
+    meso assignments [n], fine counts per meso cluster)."""
+    if kind == "f32":
+        X = _c(data, np.float32)
+        n = X.shape[0]
+        Cm, am, _ = lloyd_f32(X, X[meso_init], meso_iters)
+    elif kind == "sq8":
+        X = _c(data, np.uint8)
+        n = X.shape[0]
+        Cm, am = lloyd_sq8(X, X[meso_init], meso_iters)
+    else:
+        r = data
+        n = r["codes"].shape[0]
+        C0 = rbq1_decode_points(r["codes"], r["F"], r["d"], r["m"], r["e"], meso_init)
+        Cm, am = lloyd_rbq1(r["codes"], r["nx2"], r["F"], r["popx"], r["d"], r["m"], C0, meso_iters, r["e"])
+    sizes = np.bincount(am, minlength=m)
+    kf = fine_counts(sizes, k)
+    base = np.concatenate([[0], np.cumsum(kf)]).astype(np.int64)
+    a = np.empty(n, np.int32)
+    Cs = []
+    for i in range(m):
+        members = np.nonzero(am == i)[0]  # increasing point index
+        if kf[i] == 0:
+            continue
+        pos = fine_init_positions(len(members), kf[i])
+        init = members[pos]
+        if kind == "f32":
+            Ci, ai, _ = lloyd_f32(X[members], X[init], fine_iters)
+        elif kind == "sq8":
+            Ci, ai = lloyd_sq8(X[members], X[init], fine_iters)
+        else:
+            C0 = rbq1_decode_points(r["codes"], r["F"], r["d"], r["m"], r["e"], init)
+            Ci, ai = lloyd_rbq1(r["codes"][members], r["nx2"][members], r["F"][members], r["popx"][members],
+                                r["d"], r["m"], C0, fine_iters, r["e"])
+        Cs.append(Ci)
+        a[members] = ai + base[i]
+    C = np.concatenate(Cs, axis=0)
+    if refine:  # one vanilla iteration over all points, then the final assignment
+        if kind == "f32":
+            C, a, _ = lloyd_f32(X, C, 1)
+        elif kind == "sq8":
+            C, a = lloyd_sq8(X, C, 1)
+        else:
+            C, a = lloyd_rbq1(r["codes"], r["nx2"], r["F"], r["popx"], r["d"], r["m"], C, 1, r["e"])
+    return C, a, am, kf

@@ -104,6 +104,15 @@ struct TcParams {
     const float *F;
     const int32_t *popx;
     int d;
+    // Segmented mode (all NULL otherwise): the point rows are sorted by
+    // group and row r may only take centroids [seg_base[g], seg_base[g + 1])
+    // of its group g = seg_group[r]; point tile rt covers the centroid tiles
+    // seg_ct0[rt] .. seg_ct0[rt] + seg_nct[rt] - 1.
+    const int32_t *seg_ct0;
+    const int32_t *seg_nct;
+    const int32_t *seg_group;
+    const int32_t *seg_base;
+    int nseg;
 };
 
 // ------------------------------------------------------------- PTX helpers
@@ -358,7 +367,23 @@ __device__ __forceinline__ void screen_insert(ScreenRow &s, float L, int j) {
     }
 }
 
-template <int MODE, int NH, int CL>
+// Centroid tiles [lo, hi) of point tile rt (every tile, or the tile's
+// groups' range in segmented mode; none past the last point tile there).
+__device__ __forceinline__ void ct_range(const TcParams &p, int64_t rt, int &lo, int &hi) {
+    if (p.seg_ct0) {
+        if (rt < p.nrt) {
+            lo = p.seg_ct0[rt];
+            hi = lo + p.seg_nct[rt];
+        } else {
+            lo = hi = 0;
+        }
+    } else {
+        lo = 0;
+        hi = p.nct;
+    }
+}
+
+template <int MODE, int NH, int CL, bool SEG>
 __global__ void __launch_bounds__(tc_threads<NH>(), 1)
     tc_assign_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                      const TcParams p) {
@@ -423,7 +448,9 @@ __global__ void __launch_bounds__(tc_threads<NH>(), 1)
             uint32_t it = 0;
             for (int64_t g = g0; g < ngroups; g += gstep) {
                 const int64_t rt = g * CL + crank;
-                for (int ct = 0; ct < p.nct; ++ct)
+                int ct_lo, ct_hi;
+                ct_range(p, rt, ct_lo, ct_hi);
+                for (int ct = ct_lo; ct < ct_hi; ++ct)
                     for (int kc = 0; kc < p.nkc; ++kc, ++it) {
                         const uint32_t s = it % STAGES, ph = (it / STAGES) & 1u;
                         if (!mbar_wait(empty_bar(s), ph ^ 1u, abort_flag)) goto producer_done;
@@ -442,8 +469,10 @@ __global__ void __launch_bounds__(tc_threads<NH>(), 1)
     } else if (warp == 1) {
         if (lane == 0) {  // ---------------------------------------- MMA issuer
             uint32_t it = 0, job = 0;
-            for (int64_t g = g0; g < ngroups; g += gstep)
-                for (int ct = 0; ct < p.nct; ++ct, ++job) {
+            for (int64_t g = g0; g < ngroups; g += gstep) {
+                int ct_lo, ct_hi;
+                ct_range(p, g * CL + crank, ct_lo, ct_hi);
+                for (int ct = ct_lo; ct < ct_hi; ++ct, ++job) {
                     const uint32_t b = job & 1u, bph = (job >> 1) & 1u;
                     if (!mbar_wait(tempty_bar(b), bph ^ 1u, abort_flag)) goto mma_done;
                     tc_fence_after();
@@ -468,6 +497,7 @@ __global__ void __launch_bounds__(tc_threads<NH>(), 1)
                     }
                     tc_commit(tfull_bar(b));
                 }
+            }
         mma_done:;
         }
     } else {  // ------------------------------------------------------- epilogue
@@ -512,7 +542,11 @@ __global__ void __launch_bounds__(tc_threads<NH>(), 1)
                 if (te < 256) reinterpret_cast<int32_t *>(rb)[te] = pre1;
             }
         };
-        rec_load(0);
+        {
+            int lo0, hi0;
+            ct_range(p, g0 * CL + crank, lo0, hi0);
+            rec_load(lo0);
+        }
         // A warp whose barrier wait gave up stops computing but keeps taking part
         // in the named barriers, so the other epilogue warps never wait on it.
         bool dead = false;
@@ -527,6 +561,21 @@ __global__ void __launch_bounds__(tc_threads<NH>(), 1)
             float fbest = INFINITY;
             float a2 = 0.0f, w2 = 0.0f, rnx2 = 0.0f, rf2 = 0.0f, rpc = 0.0f;
             int32_t nxr = 0;
+            // segmented mode: this row's centroid range (ids clamped into bounds)
+            int cb = 0, ce = 0x7fffffff;
+            if (SEG && valid) {
+                int gi = p.seg_group[row];
+                gi = gi < 0 ? 0 : (gi >= p.nseg ? p.nseg - 1 : gi);
+                cb = p.seg_base[gi];
+                ce = p.seg_base[gi + 1];
+            }
+            int ct_lo, ct_hi;
+            ct_range(p, rt, ct_lo, ct_hi);
+            int next_lo = 0;
+            {
+                int nhi;
+                ct_range(p, (g + gstep) * CL + crank, next_lo, nhi);
+            }
             if (MODE == MODE_SCREEN) {
                 a2 = valid ? 2.0f * p.xinfo[row].x : 0.0f;
                 // 2 W_row, W_row = 2 ||x~|| max h' + max z >= every pair's half-width
@@ -538,14 +587,14 @@ __global__ void __launch_bounds__(tc_threads<NH>(), 1)
                 rf2 = valid ? __fmul_rn(-2.0f, p.F[row]) : 0.0f;  // exact
                 rpc = valid ? (float)(2 * p.popx[row] - p.d) : 0.0f;
             }
-            for (int ct = 0; ct < p.nct; ++ct, ++job) {
+            for (int ct = ct_lo; ct < ct_hi; ++ct, ++job) {
                 const uint32_t b = job & 1u, bph = (job >> 1) & 1u;
                 bool ok = true;
                 if (!dead) ok = mbar_wait(tfull_bar(b), bph, abort_flag);
                 dead = dead || !__all_sync(0xffffffffu, ok);
                 rec_store(b);
                 asm volatile("bar.sync 2, %0;" ::"n"(epi_threads<NH>()) : "memory");
-                rec_load(ct + 1 < p.nct ? ct + 1 : 0);
+                rec_load(ct + 1 < ct_hi ? ct + 1 : next_lo);
                 if (dead) continue;
                 tc_fence_after();
                 const uint8_t *rbuf = rec_base + b * REC_BYTES;
@@ -576,16 +625,32 @@ __global__ void __launch_bounds__(tc_threads<NH>(), 1)
                                 v[i + 1] = __float_as_uint(st.y);
                             }
                         }
+                        if (SEG && (j0 < cb || j0 + 32 > ce)) {
+                            // segmented rows whose range cuts this chunk: columns
+                            // outside it do not exist for this row
+#pragma unroll
+                            for (int g = 0; g < 4; ++g) {
+                                cm[g] = INFINITY;
+#pragma unroll
+                                for (int i = 8 * g; i < 8 * g + 8; ++i) {
+                                    const bool in = j0 + i >= cb && j0 + i < ce;
+                                    const float x = in ? __uint_as_float(v[i]) : INFINITY;
+                                    v[i] = __float_as_uint(x);
+                                    cm[g] = fminf(cm[g], x);
+                                }
+                            }
+                        }
                         sr.umin = fminf(sr.umin, fminf(fminf(cm[0], cm[1]), fminf(cm[2], cm[3])));
                         const float thr = __fadd_ru(sr.umin, w2);
                         // pass 2 (rare once the running minimum is small): pairs within
                         // 2 W_row of the running minimum of s~ could still be the nearest
-                        if (fminf(fminf(cm[0], cm[1]), fminf(cm[2], cm[3])) <= thr) {
+                        const float cmin = fminf(fminf(cm[0], cm[1]), fminf(cm[2], cm[3]));
+                        if (cmin <= thr && cmin < INFINITY) {
                             // only the 8-column groups whose minimum is inside
                             uint32_t mask = 0;
 #pragma unroll
                             for (int g = 0; g < 4; ++g) {
-                                if (cm[g] <= thr) {
+                                if (cm[g] <= thr && cm[g] < INFINITY) {
 #pragma unroll
                                     for (int i = 8 * g; i < 8 * g + 8; ++i)
                                         mask |= (__uint_as_float(v[i]) <= thr ? 1u : 0u) << i;
@@ -602,7 +667,7 @@ __global__ void __launch_bounds__(tc_threads<NH>(), 1)
                         for (int i = 0; i < 32; ++i) {
                             const int32_t dot = __float2int_rn(__uint_as_float(v[i]));
                             const int32_t dd = nxr + reinterpret_cast<const int32_t *>(rbuf)[cc + i] - 2 * dot;
-                            if (dd < best) {
+                            if (dd < best && (!SEG || (j0 + i >= cb && j0 + i < ce))) {
                                 best = dd;
                                 besti = j0 + i;
                             }
@@ -635,7 +700,11 @@ __global__ void __launch_bounds__(tc_threads<NH>(), 1)
                                 const float2 t = fmul2(make_float2(bs.x, bs.y), make_float2(rpc, rpc));
                                 const float2 u = ffma2(make_float2(bs.z, bs.w), qv, t);
                                 const float2 nn = fadd2(make_float2(rnx2, rnx2), make_float2(qn.z, qn.w));
-                                const float2 est = ffma2(make_float2(rf2, rf2), u, nn);
+                                float2 est = ffma2(make_float2(rf2, rf2), u, nn);
+                                if (SEG && (j0 < cb || j0 + 32 > ce)) {  // columns outside the row's group
+                                    if (j0 + i < cb || j0 + i >= ce) est.x = INFINITY;
+                                    if (j0 + i + 1 < cb || j0 + i + 1 >= ce) est.y = INFINITY;
+                                }
                                 if (est.x < gb[g]) {
                                     gb[g] = est.x;
                                     gi[g] = j0 + i;
@@ -1139,17 +1208,18 @@ int launch_tc(const void *xs, int64_t n, int dp, int d, const void *cs, int k, c
     constexpr int CL = TC_CL[MODE];
     constexpr size_t SMEM = tc_smem_bytes<MODE, NH>();
     static_assert(SMEM <= 227 * 1024, "shared memory per CTA");
-    auto kern = tc_assign_kernel<MODE, NH, CL>;
+    auto kern = p0.seg_group ? tc_assign_kernel<MODE, NH, CL, true> : tc_assign_kernel<MODE, NH, CL, false>;
+    const int segi = p0.seg_group ? 1 : 0;
     // per device: the attribute and the number of clusters that fit at once
     constexpr int MAXDEV = 64;
     static std::mutex mu;
-    static int cached_clusters[3][MAXDEV] = {};
+    static int cached_clusters[3][2][MAXDEV] = {};
     int dev = 0;
     SKM_CUDA_TRY(cudaGetDevice(&dev));
     int max_clusters = 0;
     {
         std::lock_guard<std::mutex> lock(mu);
-        if (dev < MAXDEV) max_clusters = cached_clusters[MODE][dev];
+        if (dev < MAXDEV) max_clusters = cached_clusters[MODE][segi][dev];
         if (max_clusters == 0) {
             SKM_CUDA_TRY(cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)SMEM));
             if (CL > 1) {
@@ -1169,7 +1239,7 @@ int launch_tc(const void *xs, int64_t n, int dp, int d, const void *cs, int k, c
                 max_clusters = device_sms();
             }
             if (max_clusters < 1) return set_error(SKM_ERR_CUDA, "no cluster of %d CTAs fits on this device", CL);
-            if (dev < MAXDEV) cached_clusters[MODE][dev] = max_clusters;
+            if (dev < MAXDEV) cached_clusters[MODE][segi][dev] = max_clusters;
         }
     }
     CUtensorMap ma, mb;

@@ -463,3 +463,51 @@ def test_hadamard_rotate_is_orthogonal_and_preserves_distances():
     T = oracle.hadamard_rotate(E, s).astype(np.float64)
     np.testing.assert_allclose(np.abs(T), 1 / np.sqrt(128), rtol=1e-7)
     np.testing.assert_allclose(T @ T.T, np.eye(128), atol=1e-6)
+
+
+# ------------------------------------------------------ hierarchical k-means
+def test_fine_counts_apportionment():
+    # proportional: 10 clusters over sizes 50/30/20 -> 5/3/2 exactly
+    assert oracle.fine_counts([50, 30, 20], 10) == [5, 3, 2]
+    # largest remainders: 7 over 5/4/1 (N=10): floors 3,2,0 remainders 5,8,7 -> +1 to 1 and 2
+    assert oracle.fine_counts([5, 4, 1], 7) == [3, 3, 1]
+    # a tiny non-empty cluster still gets one, taken from the largest
+    assert oracle.fine_counts([98, 1, 1], 3) == [1, 1, 1]
+    assert oracle.fine_counts([990, 5, 5], 10) == [8, 1, 1]
+    # empty meso clusters get none; the total is always k
+    kf = oracle.fine_counts([0, 40, 0, 60], 9)
+    assert kf[0] == 0 and kf[2] == 0 and sum(kf) == 9
+    assert oracle.fine_init_positions(10, 4) == [0, 2, 5, 7]
+
+
+def test_hierarchical_with_one_meso_cluster_is_plain_lloyd():
+    """m = 1: every point is in the single meso cluster, so the fine phase is
+    vanilla Lloyd with init at evenly spaced points."""
+    r = _rng(31)
+    X = r.standard_normal((400, 6)).astype(np.float32)
+    C, a, am, kf = oracle.hierarchical("f32", X, 5, 1, np.array([0]), 2, 4)
+    assert kf == [5] and np.all(am == 0)
+    init = np.array(oracle.fine_init_positions(400, 5))
+    Cl, al, _ = oracle.lloyd_f32(X, X[init], 4)
+    np.testing.assert_array_equal(a, al)
+    np.testing.assert_array_equal(C, Cl)
+
+
+def test_hierarchical_recovers_separated_blobs_and_refine_does_not_hurt():
+    """Four far-apart blobs of 3 sub-blobs each, m = 4 meso and k = 12 fine
+    clusters: the meso clusters find the blobs (apportioned 3 each), the fine
+    phase the sub-blobs; the refinement iteration does not raise the WCSS."""
+    r = _rng(32)
+    cent = np.array([[0, 0], [100, 0], [0, 100], [100, 100]], np.float64)
+    sub = np.array([[0, 0], [6, 0], [0, 6]], np.float64)
+    pts = [c + s + r.normal(0, 0.3, (50, 2)) for c in cent for s in sub]
+    X = np.concatenate(pts).astype(np.float32)
+    meso_init = np.array([0, 150, 300, 450])
+    C, a, am, kf = oracle.hierarchical("f32", X, 12, 4, meso_init, 3, 5)
+    assert kf == [3, 3, 3, 3]
+    labels = np.repeat(np.arange(12), 50)
+    for s in range(12):  # each sub-blob maps to a single fine cluster
+        assert len(set(a[labels == s])) == 1
+    w = oracle.objective_f32(X, C, a)
+    C2, a2, _, _ = oracle.hierarchical("f32", X, 12, 4, meso_init, 3, 5, refine=True)
+    assert oracle.objective_f32(X, C2, a2) <= w * (1 + 1e-9)
