@@ -111,7 +111,7 @@ uint64_t skm_kernel_launches(void);
 
 /* Bytes of scratch needed by op for these points and k centroids.
  * op: 0 = skm_assign, 1 = skm_update, 2 = skm_fit, 3 = skm_quantize,
- *     4 = skm_pca_fit.
+ *     4 = skm_pca_fit, 5 = skm_assign_segmented.
  * Returns 0 with skm_last_error() set when the arguments are invalid. */
 size_t skm_workspace_size(int op, const skm_data *x, int k);
 
@@ -258,6 +258,21 @@ int skm_assign(const skm_data *x, const void *C, int k, const int32_t *prev_assi
  *   No cudaMalloc, cudaFree or allocating library call is made. */
 int skm_assign_rbq1_noalloc(const skm_data *x, const float *C, int k, int32_t *assign, float *dist,
                             void *stream);
+
+/* Segmented assignment (the FINE-CLUSTERING phase of hierarchical k-means):
+ * the rows of x are sorted by group (group[n] non-decreasing, device int32 in
+ * [0, nseg)); row r takes the nearest of the centroids [base[g], base[g+1])
+ * of its group g = group[r] only (base: device int32[nseg + 1], base[0] = 0,
+ * non-decreasing, base[nseg] <= k, every group referenced by a row non-empty),
+ * with the same per-representation rules as skm_assign (F32/BF16 exact fp32
+ * argmin; SQ8 and RBQ1 bit-exact), ties to the lowest index.  Tensor-core
+ * paths only: SQ8 and RBQ1 need d <= 1024; no pruning flag.  Group ids
+ * outside [0, nseg) are clamped (never an out-of-bounds access); unsorted
+ * groups give undefined assignments.  Workspace: skm_workspace_size(5, x, k).
+ * Asynchronous. */
+int skm_assign_segmented(const skm_data *x, const void *C, int k, const int32_t *group,
+                         const int32_t *base, int nseg, int32_t *assign, float *dist, void *ws,
+                         size_t ws_bytes, void *stream);
 
 /* ------------------------------------------------------------------------
  * Update, Section 2.3 STEP 3 (and the quantized-domain variants of 3.1).

@@ -26,7 +26,7 @@ REPR_F32, REPR_SQ8, REPR_RBQ1, REPR_BF16 = 0, 1, 2, 3
 FLAG_PRUNE = 1
 DTYPE_F32, DTYPE_BF16 = 0, 1
 EMPTY_KEEP, EMPTY_SPLIT = 0, 1
-OP_ASSIGN, OP_UPDATE, OP_FIT, OP_QUANTIZE, OP_PCA = 0, 1, 2, 3, 4
+OP_ASSIGN, OP_UPDATE, OP_FIT, OP_QUANTIZE, OP_PCA, OP_ASSIGN_SEG = 0, 1, 2, 3, 4, 5
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
 _LIB_PATH = os.path.join(_HERE, "_build", "libskm.so")
@@ -37,6 +37,7 @@ EXPORTED_SYMBOLS = [
     "skm_last_error", "skm_version", "skm_kernel_launches", "skm_workspace_size", "skm_screen_bytes",
     "skm_screen_prep", "skm_project", "skm_project_hadamard", "skm_make_rotation",
     "skm_pca_fit", "skm_quantize", "skm_rbq1_exponent", "skm_assign", "skm_assign_rbq1_noalloc",
+    "skm_assign_segmented",
     "skm_update",
     "skm_merge_partials", "skm_update_finalize", "skm_fit", "skm_split_empty", "skm_objective",
     "skm_sq8_decode",
@@ -106,6 +107,7 @@ def lib():
             "skm_rbq1_exponent": ([vp, i64, vp, vp, sz, vp], i32),
             "skm_assign": ([vp, vp, i32, vp, vp, vp, vp, sz, vp], i32),
             "skm_assign_rbq1_noalloc": ([vp, vp, i32, vp, vp, vp], i32),
+            "skm_assign_segmented": ([vp, vp, i32, vp, vp, i32, vp, vp, vp, sz, vp], i32),
             "skm_update": ([vp, vp, i32, vp, vp, vp, vp, sz, vp], i32),
             "skm_merge_partials": ([vp, vp, i64, i32, vp], i32),
             "skm_update_finalize": ([vp, vp, vp, i32, vp, vp], i32),
@@ -311,6 +313,20 @@ def skm_assign_rbq1_noalloc(pts: Points, C, out, dist_out=None, stream=None):
     _check(lib().skm_assign_rbq1_noalloc(ctypes.byref(pts.ref), _ptr(C), C.shape[0], _ptr(out), _ptr(dist_out),
                                          _stream(stream)))
     return out, dist_out
+
+
+def skm_assign_segmented(pts: Points, C, group, base, want_dist=True, ws=None, stream=None, out=None):
+    """Rows sorted by group; row r takes the nearest of C[base[g]:base[g+1]], g = group[r]."""
+    k = C.shape[0]
+    dev = pts.device
+    if ws is None:
+        ws = _ws(skm_workspace_size(OP_ASSIGN_SEG, pts, k), dev)
+    assign = out if out is not None else torch.empty(pts.n, device=dev, dtype=torch.int32)
+    dist = torch.empty(pts.n, device=dev, dtype=torch.float32) if want_dist else None
+    _check(lib().skm_assign_segmented(ctypes.byref(pts.ref), _ptr(C), int(k), _ptr(group), _ptr(base),
+                                      int(base.numel() - 1), _ptr(assign), _ptr(dist), _ptr(ws), ws.numel(),
+                                      _stream(stream)))
+    return assign, dist
 
 
 def skm_update(pts: Points, assign, C_inout, counts=None, partial=None, ws=None, stream=None):

@@ -1160,6 +1160,69 @@ __global__ void add_stats_kernel(const int32_t *__restrict__ counters, int64_t *
     stats[2] |= counters[2];
 }
 
+// ---------------------------------------------------------- segmented mode
+// Centroid tiles of each point tile: the union of its rows' group ranges
+// (min and max group over the tile's rows, ids clamped into [0, nseg)).
+__global__ void seg_tiles_kernel(const int32_t *__restrict__ group, const int32_t *__restrict__ base, int nseg,
+                                 int64_t n, int64_t nrt, int32_t *__restrict__ ct0, int32_t *__restrict__ nct) {
+    const int lane = threadIdx.x & 31;
+    const int64_t warp = (blockIdx.x * (int64_t)blockDim.x + threadIdx.x) >> 5;
+    const int64_t nw = ((int64_t)gridDim.x * blockDim.x) >> 5;
+    for (int64_t rt = warp; rt < nrt; rt += nw) {
+        int gmin = 0x7fffffff, gmax = -1;
+        for (int i = lane; i < BM; i += 32) {
+            const int64_t r = rt * BM + i;
+            if (r < n) {
+                int g = group[r];
+                g = g < 0 ? 0 : (g >= nseg ? nseg - 1 : g);
+                gmin = min(gmin, g);
+                gmax = max(gmax, g);
+            }
+        }
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) {
+            gmin = min(gmin, __shfl_xor_sync(0xffffffffu, gmin, o));
+            gmax = max(gmax, __shfl_xor_sync(0xffffffffu, gmax, o));
+        }
+        if (lane == 0) {
+            const int lo = base[gmin], hi = base[gmax + 1];
+            const int t0 = lo / BN;
+            const int t1 = hi > lo ? (hi + BN - 1) / BN : t0 + 1;
+            ct0[rt] = t0;
+            nct[rt] = t1 - t0;
+        }
+    }
+}
+
+// Segmented fallback: one warp per listed row scans its own group's range in
+// fp32 (direct differences), ties to the lowest index.
+template <typename TX>
+__global__ void seg_rows_exact_kernel(const TX *__restrict__ X, int d, const float *__restrict__ C,
+                                      const int32_t *__restrict__ rows, const int32_t *__restrict__ count,
+                                      const int32_t *__restrict__ group, const int32_t *__restrict__ base,
+                                      int nseg, int32_t *__restrict__ assign) {
+    const int lane = threadIdx.x & 31;
+    const int64_t warp = (blockIdx.x * (int64_t)blockDim.x + threadIdx.x) >> 5;
+    const int64_t nw = ((int64_t)gridDim.x * blockDim.x) >> 5;
+    const int64_t cnt = *count;
+    for (int64_t t = warp; t < cnt; t += nw) {
+        const int64_t r = rows[t];
+        int g = group[r];
+        g = g < 0 ? 0 : (g >= nseg ? nseg - 1 : g);
+        const int cb = base[g], ce = base[g + 1];
+        float bd = INFINITY;
+        int bj = cb;
+        for (int j = cb; j < ce; ++j) {
+            const float dd = warp_sqdist<TX>(X + r * d, C + (int64_t)j * d, d, lane);
+            if (dd < bd) {
+                bd = dd;
+                bj = j;
+            }
+        }
+        if (lane == 0) assign[r] = bj;
+    }
+}
+
 // ------------------------------------------------------------------ host side
 PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
     static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
@@ -1423,8 +1486,25 @@ int tc_init_stats(TcAssignBufs &b, cudaStream_t st) {
     return SKM_OK;
 }
 
+// point tiles' centroid-tile ranges for a segmented call (none otherwise)
+static int seg_setup(const TcSeg *seg, int64_t n, TcParams &p, cudaStream_t st) {
+    if (!seg) return SKM_OK;
+    const int64_t nrt = cdiv(n, BM);
+    int64_t blocks = (nrt * 32 + 255) / 256;
+    if (blocks > 152 * 8) blocks = 152 * 8;
+    seg_tiles_kernel<<<(int)(blocks < 1 ? 1 : blocks), 256, 0, st>>>(seg->group, seg->base, seg->nseg, n, nrt,
+                                                                    seg->ct0, seg->nct);
+    SKM_CUDA_TRY(launched());
+    p.seg_ct0 = seg->ct0;
+    p.seg_nct = seg->nct;
+    p.seg_group = seg->group;
+    p.seg_base = seg->base;
+    p.nseg = seg->nseg;
+    return SKM_OK;
+}
+
 int tc_assign_float(const skm_data *x, const float *C, int k, int32_t *assign, float *dist,
-                    TcAssignBufs &b, cudaStream_t st) {
+                    TcAssignBufs &b, cudaStream_t st, const TcSeg *seg) {
     const int64_t n = x->n;
     const int d = x->d, dp = round8(d);
     const bool bf16 = x->repr == SKM_REPR_BF16;
@@ -1454,14 +1534,21 @@ int tc_assign_float(const skm_data *x, const float *C, int k, int32_t *assign, f
     p.fall_rows = b.fall_rows;
     p.counters = b.counters;
     p.assign = assign;
+    SKM_TRY(seg_setup(seg, n, p, st));
     SKM_TRY(launch_tc<MODE_SCREEN>(v.xs, n, dp, d, b.cs, k, p, st));
     const int gw = grid_warps(n);
     if (bf16) {
         const uint16_t *X = static_cast<const uint16_t *>(x->x);
         rescore_kernel<uint16_t><<<gw, 256, 0, st>>>(X, d, C, b.resc_rows, b.counters, b.cand, assign);
         SKM_CUDA_TRY(launched());
-        SKM_CUDA_TRY(launch_assign_exact_rows(X, 1, b.fall_rows, b.counters + 1, n, d, C, k, assign,
-                                              nullptr, b.fall_keys, st));
+        if (seg) {
+            seg_rows_exact_kernel<uint16_t><<<gw, 256, 0, st>>>(X, d, C, b.fall_rows, b.counters + 1, seg->group,
+                                                                seg->base, seg->nseg, assign);
+            SKM_CUDA_TRY(launched());
+        } else {
+            SKM_CUDA_TRY(launch_assign_exact_rows(X, 1, b.fall_rows, b.counters + 1, n, d, C, k, assign,
+                                                  nullptr, b.fall_keys, st));
+        }
         if (dist) {
             assigned_dist_kernel<uint16_t><<<gw, 256, 0, st>>>(X, n, d, C, assign, dist);
             SKM_CUDA_TRY(launched());
@@ -1470,8 +1557,14 @@ int tc_assign_float(const skm_data *x, const float *C, int k, int32_t *assign, f
         const float *X = static_cast<const float *>(x->x);
         rescore_kernel<float><<<gw, 256, 0, st>>>(X, d, C, b.resc_rows, b.counters, b.cand, assign);
         SKM_CUDA_TRY(launched());
-        SKM_CUDA_TRY(launch_assign_exact_rows(X, 0, b.fall_rows, b.counters + 1, n, d, C, k, assign,
-                                              nullptr, b.fall_keys, st));
+        if (seg) {
+            seg_rows_exact_kernel<float><<<gw, 256, 0, st>>>(X, d, C, b.fall_rows, b.counters + 1, seg->group,
+                                                             seg->base, seg->nseg, assign);
+            SKM_CUDA_TRY(launched());
+        } else {
+            SKM_CUDA_TRY(launch_assign_exact_rows(X, 0, b.fall_rows, b.counters + 1, n, d, C, k, assign,
+                                                  nullptr, b.fall_keys, st));
+        }
         if (dist) {
             assigned_dist_kernel<float><<<gw, 256, 0, st>>>(X, n, d, C, assign, dist);
             SKM_CUDA_TRY(launched());
@@ -1484,10 +1577,11 @@ int tc_assign_float(const skm_data *x, const float *C, int k, int32_t *assign, f
 
 int tc_assign_sq8(const skm_data *x, const uint8_t *C, int k, int32_t *nx_plain,
                   int32_t *nc_plain, int32_t *assign, float *dist, TcAssignBufs &b,
-                  cudaStream_t st) {
+                  cudaStream_t st, const TcSeg *seg) {
     const int64_t n = x->n;
     const int d = x->d, dp = round8(d);
     if (d > TC_SQ8_MAX_D) {  // the bf16 accumulation is exact only up to d = 1024
+        if (seg) return set_error(SKM_ERR_UNSUPPORTED, "segmented SQ8 assignment needs d <= %d", TC_SQ8_MAX_D);
         const uint8_t *X = static_cast<const uint8_t *>(x->x);
         SKM_CUDA_TRY(launch_row_sqnorm_u8(X, n, d, nx_plain, st));
         SKM_CUDA_TRY(launch_row_sqnorm_u8(C, k, d, nc_plain, st));
@@ -1511,6 +1605,7 @@ int tc_assign_sq8(const skm_data *x, const uint8_t *C, int k, int32_t *nx_plain,
     p.nx = v.nx;
     p.nc = b.nc;
     p.dist = dist;
+    SKM_TRY(seg_setup(seg, n, p, st));
     SKM_TRY(launch_tc<MODE_SQ8>(v.xs, n, dp, d, b.cs, k, p, st));
     add_stats_kernel<<<1, 1, 0, st>>>(b.counters, b.stats);
     SKM_CUDA_TRY(launched());
@@ -1518,7 +1613,7 @@ int tc_assign_sq8(const skm_data *x, const uint8_t *C, int k, int32_t *nx_plain,
 }
 
 int tc_assign_rbq1(const skm_data *x, const float *C, int k, int32_t *assign, float *dist,
-                   TcAssignBufs &b, cudaStream_t st) {
+                   TcAssignBufs &b, cudaStream_t st, const TcSeg *seg) {
     const int64_t n = x->n;
     const int d = x->d, dp = round16(d);
     const void *screen = x->screen;
@@ -1545,6 +1640,7 @@ int tc_assign_rbq1(const skm_data *x, const float *C, int k, int32_t *assign, fl
     p.F = x->F;
     p.popx = x->popx;
     p.d = d;
+    SKM_TRY(seg_setup(seg, n, p, st));
     SKM_TRY(launch_tc<MODE_RBQ1>(v.xs, n, dp, d, b.cs, k, p, st));
     add_stats_kernel<<<1, 1, 0, st>>>(b.counters, b.stats);
     SKM_CUDA_TRY(launched());

@@ -311,6 +311,14 @@ size_t skm_workspace_size(int op, const skm_data *x, int k) {
         plan_fit(x, k, cv, b);
         break;
     }
+    case 5: {  // segmented assignment
+        if (check_data(x, false) || check_k(x, k)) return 0;
+        AssignBufs b;
+        plan_assign(x, k, cv, b);
+        cv.take<int32_t>((size_t)cdiv(x->n, 128));
+        cv.take<int32_t>((size_t)cdiv(x->n, 128));
+        break;
+    }
     case 3: {  // quantize: column reductions
         if (!x || x->d < 1 || x->d > MAX_D) {
             set_error(SKM_ERR_INVALID_ARG, "bad skm_data for op 3");
@@ -502,6 +510,46 @@ int skm_assign(const skm_data *x, const void *C, int k, const int32_t *prev_assi
     plan_assign(x, k, cv, b);
     SKM_TRY(need_ws(cv, ws_bytes, ws));
     return do_assign(x, C, k, prev_assign, assign, dist, b, S(stream));
+}
+
+// Segmented assignment (the fine phase of hierarchical k-means): tensor-core
+// paths only; the row-tile ranges are derived on the device.
+static int do_assign_seg(const skm_data *x, const void *C, int k, const int32_t *group, const int32_t *base,
+                         int nseg, int32_t *assign, float *dist, AssignBufs &b, int32_t *ct0, int32_t *nct,
+                         cudaStream_t st) {
+    TcSeg sg;
+    sg.group = group;
+    sg.base = base;
+    sg.nseg = nseg;
+    sg.ct0 = ct0;
+    sg.nct = nct;
+    switch (x->repr) {
+    case SKM_REPR_F32:
+    case SKM_REPR_BF16:
+        return tc_assign_float(x, static_cast<const float *>(C), k, assign, dist, b.tc, st, &sg);
+    case SKM_REPR_SQ8:
+        return tc_assign_sq8(x, static_cast<const uint8_t *>(C), k, b.nx, b.nc, assign, dist, b.tc, st, &sg);
+    default:
+        if (x->d > TC_RBQ1_MAX_D)
+            return set_error(SKM_ERR_UNSUPPORTED, "segmented RBQ1 assignment needs d <= %d", TC_RBQ1_MAX_D);
+        return tc_assign_rbq1(x, static_cast<const float *>(C), k, assign, dist, b.tc, st, &sg);
+    }
+}
+
+int skm_assign_segmented(const skm_data *x, const void *C, int k, const int32_t *group, const int32_t *base,
+                         int nseg, int32_t *assign, float *dist, void *ws, size_t ws_bytes, void *stream) {
+    SKM_TRY(check_data(x));
+    SKM_TRY(check_k(x, k));
+    if (!C || !assign || !group || !base || nseg < 1)
+        return set_error(SKM_ERR_INVALID_ARG, "C, assign, group, base and nseg >= 1 are required");
+    if (use_prune(x)) return set_error(SKM_ERR_UNSUPPORTED, "segmented assignment has no pruning variant");
+    Carver cv(ws, ws_bytes);
+    AssignBufs b;
+    plan_assign(x, k, cv, b);
+    int32_t *ct0 = cv.take<int32_t>((size_t)cdiv(x->n, 128));
+    int32_t *nct = cv.take<int32_t>((size_t)cdiv(x->n, 128));
+    SKM_TRY(need_ws(cv, ws_bytes, ws));
+    return do_assign_seg(x, C, k, group, base, nseg, assign, dist, b, ct0, nct, S(stream));
 }
 
 int skm_update(const skm_data *x, const int32_t *assign, int k, void *C_inout, int64_t *counts,

@@ -30,21 +30,32 @@ struct TcAssignBufs {
     unsigned long long *fall_keys = nullptr;  // F32/BF16: per fallback row, (dist bits, index)
 };
 
+// Segmented assignment: rows sorted by group, row r only takes centroids
+// [base[g], base[g + 1]) of g = group[r]; ct0 / nct: workspace of one int32
+// per 128-row point tile.
+struct TcSeg {
+    const int32_t *group = nullptr;
+    const int32_t *base = nullptr;
+    int nseg = 0;
+    int32_t *ct0 = nullptr;
+    int32_t *nct = nullptr;
+};
+
 size_t tc_screen_bytes(int repr, int64_t n, int d, const void *x);
 int tc_screen_prep(const skm_data *x, void *screen, cudaStream_t st);
 void tc_plan(int repr, int64_t n, int d, int k, const void *x, const void *screen, Carver &cv,
              TcAssignBufs &b);
 int tc_init_stats(TcAssignBufs &b, cudaStream_t st);
 int tc_assign_float(const skm_data *x, const float *C, int k, int32_t *assign, float *dist,
-                    TcAssignBufs &b, cudaStream_t st);
+                    TcAssignBufs &b, cudaStream_t st, const TcSeg *seg = nullptr);
 // nx_plain / nc_plain: buffers for the __dp4a path (d > TC_SQ8_MAX_D), filled here.
 int tc_assign_sq8(const skm_data *x, const uint8_t *C, int k, int32_t *nx_plain,
                   int32_t *nc_plain, int32_t *assign, float *dist, TcAssignBufs &b,
-                  cudaStream_t st);
+                  cudaStream_t st, const TcSeg *seg = nullptr);
 // RBQ1 on tensor cores (e4m3 operands, exact integer P, same fp32 epilogue
 // as the AND+popcount kernel).
 int tc_assign_rbq1(const skm_data *x, const float *C, int k, int32_t *assign, float *dist,
-                   TcAssignBufs &b, cudaStream_t st);
+                   TcAssignBufs &b, cudaStream_t st, const TcSeg *seg = nullptr);
 // Copies the cumulative statistics; returns SKM_ERR_TIMEOUT if a pipeline
 // wait gave up.  Synchronises the stream.
 int tc_read_stats(const TcAssignBufs &b, skm_stats *st_host, cudaStream_t st);

@@ -563,3 +563,63 @@ def test_project_hadamard_vs_oracle(skm, n, d, D):
     Yb = skm.skm_project_hadamard(X.to(DEV), sigma.to(DEV), None if mean is None else mean.to(DEV),
                                   out_dtype=skm.DTYPE_BF16).float().cpu().numpy()
     assert np.all(np.abs(Yb - Yo) <= 2.0 ** -8 * np.abs(Yo) + 1e-6)
+
+
+# ------------------------------------------------------- segmented assignment
+_SEG_SIZES = [1, 127, 129, 300, 5, 1000, 64, 257, 2, 700]
+_SEG_KS = [1, 3, 200, 2, 40, 300, 7, 1, 2, 90]
+
+
+def _segments():
+    group = np.repeat(np.arange(len(_SEG_SIZES)), _SEG_SIZES).astype(np.int32)
+    base = np.concatenate([[0], np.cumsum(_SEG_KS)]).astype(np.int32)
+    return group, base
+
+
+@pytest.mark.parametrize("kind", ["f32", "bf16", "sq8", "rbq1"])
+def test_assign_segmented_vs_oracle_per_group(skm, kind):
+    group, base = _segments()
+    n, k, d = group.size, int(base[-1]), 96
+    X = _points(n, d, seed=41)
+    g = torch.from_numpy(group).to(DEV)
+    bt = torch.from_numpy(base).to(DEV)
+    Cf = _points(k, d, seed=42)
+    if kind in ("f32", "bf16"):
+        if kind == "bf16":
+            Xb = X.to(torch.bfloat16)
+            xb = Xb.view(torch.int16).numpy().view(np.uint16)
+            pts = skm.Points(skm.REPR_BF16, Xb.view(torch.int16).to(DEV), d)
+        else:
+            pts = skm.Points(skm.REPR_F32, X.to(DEV), d)
+        a, dist = skm.skm_assign_segmented(pts, Cf.to(DEV), g, bt)
+        ag = a.cpu().numpy()
+        for s in range(len(_SEG_SIZES)):
+            rows = np.nonzero(group == s)[0]
+            Cs = Cf.numpy()[base[s]:base[s + 1]]
+            if kind == "bf16":
+                ao, best, second = oracle.assign_bf16(xb[rows], Cs)
+            else:
+                ao, best, second = oracle.assign_f32(X.numpy()[rows], Cs)
+            _check_f32(ag[rows] - base[s], dist.cpu().numpy()[rows], best, second, ao, f"segment {s}")
+    elif kind == "sq8":
+        q = skm.skm_quantize(skm.REPR_SQ8, X.to(DEV))
+        codes = q["codes"].cpu().numpy()
+        Cc = torch.from_numpy(np.random.default_rng(43).integers(0, 256, (k, d)).astype(np.uint8))
+        pts = skm.Points(skm.REPR_SQ8, q["codes"], d)
+        a, dist = skm.skm_assign_segmented(pts, Cc.to(DEV), g, bt)
+        for s in range(len(_SEG_SIZES)):
+            rows = np.nonzero(group == s)[0]
+            ao, bo = oracle.assign_sq8(codes[rows], Cc.numpy()[base[s]:base[s + 1]])
+            np.testing.assert_array_equal(a.cpu().numpy()[rows] - base[s], ao)
+            np.testing.assert_array_equal(dist.cpu().numpy()[rows], bo.astype(np.float32))
+    else:
+        r = skm.skm_quantize(skm.REPR_RBQ1, X.to(DEV))
+        pts = skm.rbq1_points(r, d)
+        h = _rbq1_host(r)
+        a, est = skm.skm_assign_segmented(pts, Cf.to(DEV), g, bt)
+        for s in range(len(_SEG_SIZES)):
+            rows = np.nonzero(group == s)[0]
+            prep = oracle.rbq1_centroid_sq4(Cf.numpy()[base[s]:base[s + 1]], h["m"])
+            ao, eo = oracle.rbq1_assign(h["codes"][rows], h["nx2"][rows], h["F"][rows], h["popx"][rows], d, prep)
+            np.testing.assert_array_equal(a.cpu().numpy()[rows] - base[s], ao)
+            np.testing.assert_array_equal(est.cpu().numpy()[rows], eo)
