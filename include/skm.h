@@ -336,6 +336,43 @@ int skm_fit(const skm_fit_config *cfg, const skm_data *x, const void *C_init,
             double *objective_host, skm_stats *stats_host, void *ws, size_t ws_bytes,
             void *stream);
 
+/* ------------------------------------------------------------------------
+ * Hierarchical k-means (Section 4, "Other Accelerators": Hierarchical k-Means): MESO-CLUSTERING
+ * of all points into m clusters (Lloyd, `meso_iters` iterations, Forgy
+ * initial centroids meso_init_idx[0..m), device int64), then FINE-CLUSTERING
+ * inside every meso cluster at once: meso cluster i gets k_i of the k fine
+ * clusters, k apportioned by the meso sizes n_i (floor of k n_i / N, the
+ * rest to the largest remainders k n_i mod N, ties to the lower index; a
+ * non-empty meso cluster left with none takes one from the one with the
+ * most; the paper states sqrt(n_i) per meso cluster, this keeps the total at
+ * k), initial fine centroids the members at positions floor(t n_i / k_i),
+ * t < k_i, in increasing point order, and `fine_iters` Lloyd iterations in
+ * which a point only takes its own meso cluster's fine centroids, then a
+ * final such assignment.  refine != 0 adds the optional vanilla iteration
+ * over all points and all k centroids, then a final vanilla assignment.
+ * Fine centroids of meso cluster i are rows sum_{j<i} k_j .. + k_i - 1.
+ *  Representations: F32, SQ8 and RBQ1 (SQ8 / RBQ1 with d <= 1024); no
+ *  pruning flag.  m <= min(k, 12288); k <= n.
+ *  Outputs (device): C_out (k rows, per-repr layout of skm_assign),
+ *  assign_out int32[n]; optional meso_assign_out int32[n] (device) and
+ *  fine_counts_host int32[m] (host); stats_host may be NULL.
+ *  Workspace: skm_hier_workspace_size (it holds a copy of the points in meso
+ *  order).  Synchronises `stream`. */
+typedef struct skm_hier_config {
+    int32_t k;
+    int32_t m;
+    int32_t meso_iters;
+    int32_t fine_iters;
+    int32_t refine;
+    int32_t reserved[3];
+} skm_hier_config;
+
+size_t skm_hier_workspace_size(const skm_hier_config *cfg, const skm_data *x);
+int skm_fit_hierarchical(const skm_hier_config *cfg, const skm_data *x, const int64_t *meso_init_idx,
+                         void *C_out, int32_t *assign_out, int32_t *meso_assign_out,
+                         int32_t *fine_counts_host, skm_stats *stats_host, void *ws, size_t ws_bytes,
+                         void *stream);
+
 /* Split large clusters into the empty ones (the library's reading of
  * Section 2.3 STEP 3).  Clusters with counts[j] == 0, in increasing j, each
  * take the current largest cluster L (most members, ties to the lowest

@@ -39,8 +39,8 @@ EXPORTED_SYMBOLS = [
     "skm_pca_fit", "skm_quantize", "skm_rbq1_exponent", "skm_assign", "skm_assign_rbq1_noalloc",
     "skm_assign_segmented",
     "skm_update",
-    "skm_merge_partials", "skm_update_finalize", "skm_fit", "skm_split_empty", "skm_objective",
-    "skm_sq8_decode",
+    "skm_merge_partials", "skm_update_finalize", "skm_fit", "skm_split_empty", "skm_hier_workspace_size",
+    "skm_fit_hierarchical", "skm_objective", "skm_sq8_decode",
 ]
 
 
@@ -73,6 +73,11 @@ class Stats(ctypes.Structure):
     _fields_ = [("rescored_rows", ctypes.c_int64), ("fallback_rows", ctypes.c_int64),
                 ("empty_clusters", ctypes.c_int64), ("prune_first_block", ctypes.c_int64),
                 ("prune_complete", ctypes.c_int64), ("reserved", ctypes.c_int64 * 3)]
+
+
+class HierConfig(ctypes.Structure):
+    _fields_ = [("k", ctypes.c_int32), ("m", ctypes.c_int32), ("meso_iters", ctypes.c_int32),
+                ("fine_iters", ctypes.c_int32), ("refine", ctypes.c_int32), ("reserved", ctypes.c_int32 * 3)]
 
 
 class FitConfig(ctypes.Structure):
@@ -113,6 +118,8 @@ def lib():
             "skm_update_finalize": ([vp, vp, vp, i32, vp, vp], i32),
             "skm_fit": ([vp, vp, vp, vp, vp, vp, vp, vp, vp, vp, sz, vp], i32),
             "skm_split_empty": ([vp, vp, vp, i32, vp, sz, vp], i32),
+            "skm_hier_workspace_size": ([vp, vp], sz),
+            "skm_fit_hierarchical": ([vp, vp, vp, vp, vp, vp, vp, vp, vp, sz, vp], i32),
             "skm_objective": ([vp, i32, i64, i32, vp, i32, vp, vp, vp, sz, vp], i32),
             "skm_sq8_decode": ([vp, i64, i32, vp, vp, vp, vp], i32),
         }
@@ -382,6 +389,31 @@ def skm_fit(pts: Points, k, iters, C_init=None, init_idx=None, want_objective=Tr
              "empty_clusters": st.empty_clusters, "prune_first_block": st.prune_first_block,
              "prune_complete": st.prune_complete}
     return C, assign, dist, (list(obj) if obj is not None else None), stats
+
+
+def skm_fit_hierarchical(pts: Points, k, m, meso_init_idx, meso_iters, fine_iters, refine=False, ws=None,
+                         stream=None):
+    """Returns (C [k], assign [n], meso assign [n], fine counts per meso cluster (list), stats dict)."""
+    dev = pts.device
+    cfg = HierConfig(int(k), int(m), int(meso_iters), int(fine_iters), int(bool(refine)))
+    if ws is None:
+        nbytes = lib().skm_hier_workspace_size(ctypes.byref(cfg), ctypes.byref(pts.ref))
+        if nbytes == 0:
+            raise SkmError(1, lib().skm_last_error().decode())
+        ws = _ws(nbytes, dev)
+    if pts.repr == REPR_SQ8:
+        C = torch.empty(k, pts.d, device=dev, dtype=torch.uint8)
+    else:
+        C = torch.empty(k, pts.d, device=dev, dtype=torch.float32)
+    assign = torch.empty(pts.n, device=dev, dtype=torch.int32)
+    meso = torch.empty(pts.n, device=dev, dtype=torch.int32)
+    kf = (ctypes.c_int32 * m)()
+    st = Stats()
+    _check(lib().skm_fit_hierarchical(ctypes.byref(cfg), ctypes.byref(pts.ref), _ptr(meso_init_idx), _ptr(C),
+                                      _ptr(assign), _ptr(meso), kf, ctypes.byref(st), _ptr(ws), ws.numel(),
+                                      _stream(stream)))
+    stats = {"rescored_rows": st.rescored_rows, "fallback_rows": st.fallback_rows}
+    return C, assign, meso, list(kf), stats
 
 
 def skm_objective(X, C, assign, stream=None):

@@ -707,3 +707,140 @@ cudaError_t launch_split_empty(void *C, int code_bytes, const int64_t *counts, i
 }
 
 }  // namespace skm
+
+namespace skm {
+
+// ---------------------------------------------------- stable sort by group
+// Rows ordered by group, increasing row index within a group (hierarchical
+// k-means' fine phase works on the meso clusters in this order, and its
+// initial fine centroids are positions inside each group).  Blocks own
+// SS_CHUNK consecutive rows: per-block group counts, a column scan over the
+// blocks, then each block (one warp, 32 rows at a time in order) places its
+// rows with __match_any_sync ranks, so the order is deterministic.
+constexpr int SS_CHUNK = 4096;
+
+static __device__ __forceinline__ int clamp_key(int g, int m) { return g < 0 ? 0 : (g >= m ? m - 1 : g); }
+
+__global__ void ss_hist_kernel(const int32_t *__restrict__ key, int64_t n, int m, int32_t *__restrict__ hist) {
+    extern __shared__ int32_t h[];
+    for (int j = threadIdx.x; j < m; j += blockDim.x) h[j] = 0;
+    __syncthreads();
+    const int64_t r0 = (int64_t)blockIdx.x * SS_CHUNK, r1 = min(n, r0 + SS_CHUNK);
+    for (int64_t r = r0 + threadIdx.x; r < r1; r += blockDim.x) atomicAdd(&h[clamp_key(key[r], m)], 1);
+    __syncthreads();
+    for (int j = threadIdx.x; j < m; j += blockDim.x) hist[(int64_t)blockIdx.x * m + j] = h[j];
+}
+
+// hist[b][j] (counts) -> first sorted position of block b's rows of group j;
+// sizes[j] = rows in group j.  One block.
+__global__ void ss_scan_kernel(int32_t *__restrict__ hist, int nblk, int m, int32_t *__restrict__ sizes) {
+    extern __shared__ int32_t goff[];
+    for (int j = threadIdx.x; j < m; j += blockDim.x) {
+        int32_t run = 0;
+        for (int b = 0; b < nblk; ++b) {
+            const int32_t t = hist[(int64_t)b * m + j];
+            hist[(int64_t)b * m + j] = run;
+            run += t;
+        }
+        sizes[j] = run;
+    }
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        int32_t run = 0;
+        for (int j = 0; j < m; ++j) {
+            goff[j] = run;
+            run += sizes[j];
+        }
+    }
+    __syncthreads();
+    for (int j = threadIdx.x; j < m; j += blockDim.x)
+        for (int b = 0; b < nblk; ++b) hist[(int64_t)b * m + j] += goff[j];
+}
+
+__global__ void ss_place_kernel(const int32_t *__restrict__ key, int64_t n, int m,
+                                const int32_t *__restrict__ starts, int32_t *__restrict__ perm,
+                                int32_t *__restrict__ skey) {
+    extern __shared__ int32_t cnt[];
+    const int lane = threadIdx.x;  // one warp
+    for (int j = lane; j < m; j += 32) cnt[j] = starts[(int64_t)blockIdx.x * m + j];
+    __syncwarp();
+    const int64_t r0 = (int64_t)blockIdx.x * SS_CHUNK, r1 = min(n, r0 + SS_CHUNK);
+    const unsigned lt = (1u << lane) - 1u;
+    for (int64_t s = r0; s < r1; s += 32) {
+        const int64_t r = s + lane;
+        const int g = r < r1 ? clamp_key(key[r], m) : -1;
+        const unsigned peers = __match_any_sync(0xffffffffu, g);
+        int pos = 0;
+        if (g >= 0) pos = cnt[g] + __popc(peers & lt);
+        __syncwarp();
+        if (g >= 0 && (peers & lt) == 0) cnt[g] += __popc(peers);  // the group's lowest lane
+        __syncwarp();
+        if (g >= 0) {
+            perm[pos] = (int32_t)r;
+            skey[pos] = g;
+        }
+    }
+}
+
+cudaError_t launch_stable_sort(const int32_t *key, int64_t n, int m, int32_t *hist, int32_t *sizes,
+                               int32_t *perm, int32_t *skey, cudaStream_t st) {
+    if (n == 0) return cudaSuccess;
+    const int nblk = (int)((n + SS_CHUNK - 1) / SS_CHUNK);
+    const size_t sm = sizeof(int32_t) * (size_t)m;
+    ss_hist_kernel<<<nblk, 256, sm, st>>>(key, n, m, hist);
+    cudaError_t e = launched();
+    if (e != cudaSuccess) return e;
+    ss_scan_kernel<<<1, 1024, sm, st>>>(hist, nblk, m, sizes);
+    e = launched();
+    if (e != cudaSuccess) return e;
+    ss_place_kernel<<<nblk, 32, sm, st>>>(key, n, m, hist, perm, skey);
+    return launched();
+}
+
+// dst row q = src row perm[q] (rowbytes per row); one warp per row
+__global__ void gather_rows_bytes_kernel(const uint8_t *__restrict__ src, int64_t rowbytes,
+                                         const int32_t *__restrict__ perm, int64_t n, uint8_t *__restrict__ dst,
+                                         int vec16) {
+    const int lane = threadIdx.x & 31;
+    const int64_t warp = (blockIdx.x * (int64_t)blockDim.x + threadIdx.x) >> 5;
+    const int64_t nw = ((int64_t)gridDim.x * blockDim.x) >> 5;
+    for (int64_t q = warp; q < n; q += nw) {
+        const uint8_t *s = src + (int64_t)perm[q] * rowbytes;
+        uint8_t *t = dst + q * rowbytes;
+        if (vec16) {
+            for (int64_t i = lane; i < rowbytes / 16; i += 32)
+                reinterpret_cast<uint4 *>(t)[i] = __ldg(reinterpret_cast<const uint4 *>(s) + i);
+        } else {
+            for (int64_t i = lane; i < rowbytes; i += 32) t[i] = s[i];
+        }
+    }
+}
+
+cudaError_t launch_gather_rows_bytes(const void *src, int64_t rowbytes, const int32_t *perm, int64_t n,
+                                     void *dst, cudaStream_t st) {
+    if (n == 0) return cudaSuccess;
+    const int vec16 = rowbytes % 16 == 0 && ((reinterpret_cast<uintptr_t>(src) | reinterpret_cast<uintptr_t>(dst)) & 15) == 0;
+    int64_t blocks = (n * 32 + 255) / 256;
+    if (blocks > 152 * 16) blocks = 152 * 16;
+    gather_rows_bytes_kernel<<<(int)blocks, 256, 0, st>>>(static_cast<const uint8_t *>(src), rowbytes, perm, n,
+                                                         static_cast<uint8_t *>(dst), vec16);
+    return launched();
+}
+
+// out[perm[q]] = in[q] (4-byte values)
+__global__ void unpermute_kernel(const int32_t *__restrict__ in, const int32_t *__restrict__ perm, int64_t n,
+                                 int32_t *__restrict__ out) {
+    for (int64_t q = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; q < n; q += (int64_t)gridDim.x * blockDim.x)
+        out[perm[q]] = in[q];
+}
+
+cudaError_t launch_unpermute(const void *in, const int32_t *perm, int64_t n, void *out, cudaStream_t st) {
+    if (n == 0) return cudaSuccess;
+    int64_t blocks = (n + 255) / 256;
+    if (blocks > 152 * 16) blocks = 152 * 16;
+    unpermute_kernel<<<(int)blocks, 256, 0, st>>>(static_cast<const int32_t *>(in), perm, n,
+                                                  static_cast<int32_t *>(out));
+    return launched();
+}
+
+}  // namespace skm

@@ -552,6 +552,228 @@ int skm_assign_segmented(const skm_data *x, const void *C, int k, const int32_t 
     return do_assign_seg(x, C, k, group, base, nseg, assign, dist, b, ct0, nct, S(stream));
 }
 
+// ------------------------------------------------------ hierarchical k-means
+static int64_t row_bytes(const skm_data *x) {
+    switch (x->repr) {
+    case SKM_REPR_F32:
+        return 4LL * x->d;
+    case SKM_REPR_SQ8:
+        return x->d;
+    case SKM_REPR_RBQ1:
+        return 4LL * words_of(x->d);
+    default:
+        return 2LL * x->d;
+    }
+}
+
+struct HierBufs {
+    uint8_t *meso_ws = nullptr;
+    size_t meso_ws_bytes = 0;
+    void *C_meso = nullptr;
+    int32_t *a_meso = nullptr;
+    int32_t *perm = nullptr, *skey = nullptr, *hist = nullptr, *sizes = nullptr, *base = nullptr;
+    uint8_t *rows = nullptr;  // the points in meso order
+    float *nx2 = nullptr, *F = nullptr;
+    int32_t *popx = nullptr;
+    uint8_t *screen = nullptr;
+    AssignBufs a;
+    int32_t *ct0 = nullptr, *nct = nullptr;
+    UpdateBufs u;
+    int32_t *a_sorted = nullptr;
+    int64_t *counts = nullptr;
+    int64_t *init_pos = nullptr;
+    int *status = nullptr;
+    unsigned int *maxbits = nullptr;
+    int *e_dev = nullptr;
+};
+
+static void plan_hier(const skm_data *x, int k, int m, Carver &cv, HierBufs &b) {
+    const int64_t n = x->n;
+    {
+        Carver mc(nullptr, 0);
+        FitBufs fb;
+        plan_fit(x, m, mc, fb);
+        b.meso_ws_bytes = mc.off;
+    }
+    b.meso_ws = cv.take<uint8_t>(b.meso_ws_bytes);
+    b.C_meso = cv.take<uint8_t>((size_t)m * (x->repr == SKM_REPR_SQ8 ? x->d : 4 * x->d));
+    b.a_meso = cv.take<int32_t>(n);
+    b.perm = cv.take<int32_t>(n);
+    b.skey = cv.take<int32_t>(n);
+    b.hist = cv.take<int32_t>((size_t)cdiv(n, 4096) * m);
+    b.sizes = cv.take<int32_t>(m);
+    b.base = cv.take<int32_t>((size_t)m + 1);
+    b.rows = cv.take<uint8_t>((size_t)(n * row_bytes(x)));
+    if (x->repr == SKM_REPR_RBQ1) {
+        b.nx2 = cv.take<float>(n);
+        b.F = cv.take<float>(n);
+        b.popx = cv.take<int32_t>(n);
+    }
+    skm_data xs = *x;
+    xs.x = b.rows;
+    const size_t sb = tc_screen_bytes(x->repr, n, x->d, b.rows ? b.rows : reinterpret_cast<const void *>(16));
+    b.screen = cv.take<uint8_t>(sb);
+    xs.screen = b.screen ? b.screen : reinterpret_cast<const void *>(1);  // measured: a screen is given
+    plan_assign(&xs, k, cv, b.a);
+    b.ct0 = cv.take<int32_t>((size_t)cdiv(n, 128));
+    b.nct = cv.take<int32_t>((size_t)cdiv(n, 128));
+    plan_update(&xs, k, cv, b.u);
+    b.a_sorted = cv.take<int32_t>(n);
+    b.counts = cv.take<int64_t>(k);
+    b.init_pos = cv.take<int64_t>(k);
+    b.status = cv.take<int>(1);
+    b.maxbits = cv.take<unsigned int>(1);
+    b.e_dev = cv.take<int>(1);
+}
+
+static int hier_check(const skm_hier_config *cfg, const skm_data *x) {
+    if (!cfg) return set_error(SKM_ERR_INVALID_ARG, "cfg is NULL");
+    SKM_TRY(check_data(x));
+    SKM_TRY(check_k(x, cfg->k, true));
+    if (cfg->m < 1 || cfg->m > cfg->k || cfg->m > 12288)
+        return set_error(SKM_ERR_INVALID_ARG, "m = %d outside [1, min(k, 12288)]", cfg->m);
+    if (cfg->meso_iters < 0 || cfg->fine_iters < 0 || cfg->meso_iters > 100000 || cfg->fine_iters > 100000)
+        return set_error(SKM_ERR_INVALID_ARG, "bad iteration counts");
+    if (x->repr == SKM_REPR_BF16) return set_error(SKM_ERR_UNSUPPORTED, "hierarchical fit: F32, SQ8 or RBQ1 points");
+    if (use_prune(x)) return set_error(SKM_ERR_UNSUPPORTED, "hierarchical fit has no pruning variant");
+    if ((x->repr == SKM_REPR_SQ8 && x->d > TC_SQ8_MAX_D) || (x->repr == SKM_REPR_RBQ1 && x->d > TC_RBQ1_MAX_D))
+        return set_error(SKM_ERR_UNSUPPORTED, "hierarchical SQ8 / RBQ1 fit needs d <= 1024");
+    return SKM_OK;
+}
+
+// Fine clusters per meso cluster: k apportioned by size (floor of k n_i / N,
+// the rest to the largest remainders k n_i mod N, ties to the lower index);
+// a non-empty meso cluster left with none takes one from the largest.
+static void fine_counts(const std::vector<int32_t> &sizes, int k, std::vector<int> &kf) {
+    const int m = (int)sizes.size();
+    int64_t N = 0;
+    for (int v : sizes) N += v;
+    kf.assign(m, 0);
+    std::vector<int64_t> rem(m);
+    int given = 0;
+    for (int i = 0; i < m; ++i) {
+        kf[i] = (int)((int64_t)k * sizes[i] / N);
+        rem[i] = (int64_t)k * sizes[i] % N;
+        given += kf[i];
+    }
+    std::vector<int> order(m);
+    for (int i = 0; i < m; ++i) order[i] = i;
+    std::stable_sort(order.begin(), order.end(), [&](int a, int b) { return rem[a] > rem[b]; });
+    for (int t = 0; t < k - given; ++t) kf[order[t]] += 1;
+    for (int i = 0; i < m; ++i)
+        if (sizes[i] > 0 && kf[i] == 0) {
+            int j = 0;
+            for (int t = 1; t < m; ++t)
+                if (kf[t] > kf[j]) j = t;
+            kf[j] -= 1;
+            kf[i] = 1;
+        }
+}
+
+int skm_fit_hierarchical(const skm_hier_config *cfg, const skm_data *x, const int64_t *meso_init_idx,
+                         void *C_out, int32_t *assign_out, int32_t *meso_assign_out, int32_t *fine_counts_host,
+                         skm_stats *stats_host, void *ws, size_t ws_bytes, void *stream) {
+    SKM_TRY(hier_check(cfg, x));
+    if (!meso_init_idx || !C_out || !assign_out)
+        return set_error(SKM_ERR_INVALID_ARG, "meso_init_idx, C_out and assign_out are required");
+    const int k = cfg->k, m = cfg->m;
+    const int64_t n = x->n;
+    const int d = x->d;
+    cudaStream_t st = S(stream);
+    Carver cv(ws, ws_bytes);
+    HierBufs b;
+    plan_hier(x, k, m, cv, b);
+    SKM_TRY(need_ws(cv, ws_bytes, ws));
+
+    // MESO-CLUSTERING: Lloyd with m clusters from the given Forgy indices
+    skm_fit_config mc{};
+    mc.k = m;
+    mc.iters = cfg->meso_iters;
+    SKM_TRY(skm_fit(&mc, x, nullptr, meso_init_idx, b.C_meso, b.a_meso, nullptr, nullptr, nullptr, b.meso_ws,
+                    b.meso_ws_bytes, stream));
+    if (meso_assign_out)
+        SKM_CUDA_TRY(cudaMemcpyAsync(meso_assign_out, b.a_meso, sizeof(int32_t) * n, cudaMemcpyDeviceToDevice, st));
+
+    // points in meso order (stable), fine-cluster budget per meso cluster
+    SKM_CUDA_TRY(launch_stable_sort(b.a_meso, n, m, b.hist, b.sizes, b.perm, b.skey, st));
+    std::vector<int32_t> sizes(m);
+    SKM_CUDA_TRY(cudaMemcpyAsync(sizes.data(), b.sizes, sizeof(int32_t) * m, cudaMemcpyDeviceToHost, st));
+    SKM_CUDA_TRY(cudaStreamSynchronize(st));
+    std::vector<int> kf;
+    fine_counts(sizes, k, kf);
+    std::vector<int32_t> base(m + 1, 0);
+    std::vector<int64_t> init(k);
+    int64_t off = 0;
+    for (int i = 0; i < m; ++i) {
+        base[i + 1] = base[i] + kf[i];
+        for (int t = 0; t < kf[i]; ++t) init[base[i] + t] = off + (int64_t)t * sizes[i] / kf[i];
+        off += sizes[i];
+    }
+    if (fine_counts_host)
+        for (int i = 0; i < m; ++i) fine_counts_host[i] = kf[i];
+    SKM_CUDA_TRY(cudaMemcpyAsync(b.base, base.data(), sizeof(int32_t) * (m + 1), cudaMemcpyHostToDevice, st));
+    SKM_CUDA_TRY(cudaMemcpyAsync(b.init_pos, init.data(), sizeof(int64_t) * k, cudaMemcpyHostToDevice, st));
+    SKM_CUDA_TRY(launch_gather_rows_bytes(x->x, row_bytes(x), b.perm, n, b.rows, st));
+    skm_data xs = *x;
+    xs.x = b.rows;
+    xs.screen = nullptr;
+    if (x->repr == SKM_REPR_RBQ1) {
+        SKM_CUDA_TRY(launch_gather_rows_bytes(x->nx2, 4, b.perm, n, b.nx2, st));
+        SKM_CUDA_TRY(launch_gather_rows_bytes(x->F, 4, b.perm, n, b.F, st));
+        SKM_CUDA_TRY(launch_gather_rows_bytes(x->popx, 4, b.perm, n, b.popx, st));
+        xs.nx2 = b.nx2;
+        xs.F = b.F;
+        xs.popx = b.popx;
+        SKM_CUDA_TRY(launch_rbq1_exponent(x->F, n, b.maxbits, b.e_dev, st));
+        int e = 0;
+        SKM_CUDA_TRY(cudaMemcpyAsync(&e, b.e_dev, sizeof(int), cudaMemcpyDeviceToHost, st));
+        SKM_CUDA_TRY(cudaStreamSynchronize(st));
+        xs.rbq1_exp = e;
+    }
+    SKM_TRY(tc_screen_prep(&xs, b.screen, st));
+    xs.screen = b.screen;
+    SKM_TRY(tc_init_stats(b.a.tc, st));
+
+    // FINE-CLUSTERING: every meso cluster at once, each point against its own
+    // meso cluster's fine centroids; initial centroids at evenly spaced members
+    SKM_CUDA_TRY(cudaMemsetAsync(b.status, 0, sizeof(int), st));
+    if (x->repr == SKM_REPR_RBQ1)
+        SKM_CUDA_TRY(launch_rbq1_decode_rows(static_cast<const uint32_t *>(xs.x), xs.F, n, d, x->m, xs.rbq1_exp,
+                                             b.init_pos, k, static_cast<float *>(C_out), b.status, st));
+    else
+        SKM_CUDA_TRY(launch_gather_rows(xs.x, n, x->repr == SKM_REPR_SQ8 ? 1 : 4, d, b.init_pos, k, C_out,
+                                        b.status, st));
+    SKM_CUDA_TRY(cudaMemsetAsync(b.u.flag, 0, sizeof(int32_t), st));
+    for (int it = 0; it <= cfg->fine_iters; ++it) {
+        SKM_TRY(do_assign_seg(&xs, C_out, k, b.skey, b.base, m, b.a_sorted, nullptr, b.a, b.ct0, b.nct, st));
+        if (it == cfg->fine_iters) break;
+        SKM_TRY(do_update(&xs, b.a_sorted, k, C_out, b.counts, nullptr, xs.rbq1_exp, b.u, st));
+    }
+    if (cfg->refine) {  // one vanilla iteration over all points, then the final assignment
+        SKM_TRY(do_assign(&xs, C_out, k, nullptr, b.a_sorted, nullptr, b.a, st));
+        SKM_TRY(do_update(&xs, b.a_sorted, k, C_out, b.counts, nullptr, xs.rbq1_exp, b.u, st));
+        SKM_TRY(do_assign(&xs, C_out, k, nullptr, b.a_sorted, nullptr, b.a, st));
+    }
+    SKM_CUDA_TRY(launch_unpermute(b.a_sorted, b.perm, n, assign_out, st));
+    SKM_CUDA_TRY(cudaStreamSynchronize(st));
+    skm_stats local;
+    memset(&local, 0, sizeof(local));
+    SKM_TRY(tc_read_stats(b.a.tc, &local, st));
+    int32_t uflag = 0;
+    SKM_CUDA_TRY(cudaMemcpy(&uflag, b.u.flag, sizeof(uflag), cudaMemcpyDeviceToHost));
+    if (uflag) return set_error(SKM_ERR_TIMEOUT, "an update pipeline wait exceeded its limit");
+    if (stats_host) *stats_host = local;
+    return SKM_OK;
+}
+
+size_t skm_hier_workspace_size(const skm_hier_config *cfg, const skm_data *x) {
+    if (hier_check(cfg, x)) return 0;
+    Carver cv(nullptr, 0);
+    HierBufs b;
+    plan_hier(x, cfg->k, cfg->m, cv, b);
+    return cv.off;
+}
+
 int skm_update(const skm_data *x, const int32_t *assign, int k, void *C_inout, int64_t *counts,
                void *partial, void *ws, size_t ws_bytes, void *stream) {
     SKM_TRY(check_data(x));

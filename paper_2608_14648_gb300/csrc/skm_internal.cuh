@@ -158,6 +158,14 @@ bool ring_sum_sq8_ok(const void *codes, int d);
 // y = H_D diag(sigma) [x - mean; 0] / sqrt(D), D a power of two in [32, 4096]
 cudaError_t launch_hadamard(const float *X, int64_t n, int d, const float *mean, const float *sigma, int D,
                             int out_bf16, void *Y, cudaStream_t st);
+// stable sort of rows by key in [0, m) (m <= 12288): hist int32[ceil(n/4096)][m],
+// sizes int32[m]; perm[q] = row at sorted position q, skey[q] its key
+cudaError_t launch_stable_sort(const int32_t *key, int64_t n, int m, int32_t *hist, int32_t *sizes,
+                               int32_t *perm, int32_t *skey, cudaStream_t st);
+cudaError_t launch_gather_rows_bytes(const void *src, int64_t rowbytes, const int32_t *perm, int64_t n,
+                                     void *dst, cudaStream_t st);
+// out[perm[q]] = in[q] for 4-byte values
+cudaError_t launch_unpermute(const void *in, const int32_t *perm, int64_t n, void *out, cudaStream_t st);
 // empty clusters take half of the largest one (w: k int64 of workspace)
 cudaError_t launch_split_empty(void *C, int code_bytes, const int64_t *counts, int k, int d,
                                int64_t *w, cudaStream_t st);

@@ -623,3 +623,56 @@ def test_assign_segmented_vs_oracle_per_group(skm, kind):
             ao, eo = oracle.rbq1_assign(h["codes"][rows], h["nx2"][rows], h["F"][rows], h["popx"][rows], d, prep)
             np.testing.assert_array_equal(a.cpu().numpy()[rows] - base[s], ao)
             np.testing.assert_array_equal(est.cpu().numpy()[rows], eo)
+
+
+# ------------------------------------------------------ hierarchical k-means
+def _hier_points(n, d, seed):
+    return _points(n, d, seed=seed, ncomp=24)
+
+
+@pytest.mark.parametrize("refine", [False, True])
+def test_fit_hierarchical_sq8_bitexact(skm, refine):
+    n, d, k, m = 9000, 64, 60, 8
+    X = _hier_points(n, d, 51)
+    q = skm.skm_quantize(skm.REPR_SQ8, X.to(DEV))
+    codes = q["codes"].cpu().numpy()
+    idx = synth.forgy_indices(n, m, seed=51)
+    C, a, meso, kf, _ = skm.skm_fit_hierarchical(skm.Points(skm.REPR_SQ8, q["codes"], d), k, m, idx.to(DEV), 3, 4,
+                                                 refine=refine)
+    Co, ao, amo, kfo = oracle.hierarchical("sq8", codes, k, m, idx.numpy(), 3, 4, refine=refine)
+    assert kf == kfo and sum(kf) == k
+    np.testing.assert_array_equal(meso.cpu().numpy(), amo)
+    np.testing.assert_array_equal(a.cpu().numpy(), ao)
+    np.testing.assert_array_equal(C.cpu().numpy(), Co)
+
+
+def test_fit_hierarchical_rbq1_bitexact(skm):
+    n, d, k, m = 8000, 128, 48, 6
+    X = _hier_points(n, d, 52)
+    r = skm.skm_quantize(skm.REPR_RBQ1, X.to(DEV))
+    pts = skm.rbq1_points(r, d)
+    h = _rbq1_host(r)
+    idx = synth.forgy_indices(n, m, seed=52)
+    C, a, meso, kf, _ = skm.skm_fit_hierarchical(pts, k, m, idx.to(DEV), 3, 3)
+    data = {"codes": h["codes"], "nx2": h["nx2"], "F": h["F"], "popx": h["popx"], "d": d, "m": h["m"],
+            "e": pts.rbq1_exp}
+    Co, ao, amo, kfo = oracle.hierarchical("rbq1", data, k, m, idx.numpy(), 3, 3)
+    assert kf == kfo
+    np.testing.assert_array_equal(meso.cpu().numpy(), amo)
+    np.testing.assert_array_equal(a.cpu().numpy(), ao)
+    np.testing.assert_array_equal(C.cpu().numpy(), Co)
+
+
+def test_fit_hierarchical_f32_vs_oracle(skm):
+    n, d, k, m = 12000, 48, 64, 8
+    X = _hier_points(n, d, 53)
+    idx = synth.forgy_indices(n, m, seed=53)
+    C, a, meso, kf, _ = skm.skm_fit_hierarchical(skm.Points(skm.REPR_F32, X.to(DEV), d), k, m, idx.to(DEV), 3, 4,
+                                                 refine=True)
+    Co, ao, amo, kfo = oracle.hierarchical("f32", X.numpy(), k, m, idx.numpy(), 3, 4, refine=True)
+    assert (meso.cpu().numpy() == amo).mean() >= AGREE
+    if kf == kfo and (meso.cpu().numpy() == amo).all():
+        assert (a.cpu().numpy() == ao).mean() >= AGREE
+    wg = oracle.objective_f32(X.numpy(), C.cpu().numpy(), a.cpu().numpy())
+    wo = oracle.objective_f32(X.numpy(), Co, ao)
+    assert abs(wg - wo) / wo <= 1e-3
