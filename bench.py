@@ -520,6 +520,44 @@ def run_case(args):
     print(json.dumps(out))
 
 
+def _run_hier(args, name, n, k, idx, runs):
+    """Flat Lloyd (skm_fit, `iters` iterations + final assignment) against
+    hierarchical k-means (m = round(sqrt k) meso clusters, `iters` meso and
+    `iters` fine iterations + final assignments), whole calls timed with CUDA
+    events after one warm-up call each."""
+    import math
+
+    import torch
+
+    import paper_2608_14648_gb300 as skm
+
+    m = max(1, round(math.sqrt(k)))
+    midx = idx[:m].contiguous()
+    for label, pts, C, d, peak, kind in runs:
+        if label not in ("fp32", "sq8", "rbq1"):
+            continue
+        ev = [torch.cuda.Event(enable_timing=True) for _ in range(4)]
+        ws = skm.workspace(skm.OP_FIT, pts, k)
+        skm.skm_fit(pts, k, args.iters, init_idx=idx, want_objective=False, want_dist=False, ws=ws)
+        ev[0].record()
+        skm.skm_fit(pts, k, args.iters, init_idx=idx, want_objective=False, want_dist=False, ws=ws)
+        ev[1].record()
+        torch.cuda.synchronize()
+        del ws
+        skm.skm_fit_hierarchical(pts, k, m, midx, args.iters, args.iters)
+        ev[2].record()
+        _, _, _, kf, _ = skm.skm_fit_hierarchical(pts, k, m, midx, args.iters, args.iters)
+        ev[3].record()
+        torch.cuda.synchronize()
+        t_flat = ev[0].elapsed_time(ev[1])
+        t_h = ev[2].elapsed_time(ev[3])
+        out = {"config": args.config, "workload": name, "repr": label, "n": n, "d": d, "k": k, "m": m,
+               "iters": args.iters, "flat_fit_ms": round(t_flat, 3), "hierarchical_fit_ms": round(t_h, 3),
+               "speedup": round(t_flat / t_h, 2), "fine_counts_min_max": [min(kf), max(kf)]}
+        print(json.dumps(out), flush=True)
+        torch.cuda.empty_cache()
+
+
 def run_config(args):
     """One JSON line per representation of a workload configuration: the
     median over Lloyd iterations 2..iters of (centroid prep + assign + update)
@@ -575,6 +613,9 @@ def run_config(args):
         runs.append(("bf16_prune", skm.Points(skm.REPR_BF16, Yb, dp, flags=skm.FLAG_PRUNE), Cb.clone(), dp,
                      None, "fp32 CUDA cores"))
     torch.cuda.synchronize()
+    if args.hier:
+        _run_hier(args, name, n, k, idx, runs)
+        return
     for label, pts, C, d, peak, kind in runs:
         C = C.clone()
         wsA = skm.workspace(skm.OP_ASSIGN, pts, k)
@@ -635,6 +676,8 @@ def main():
     ap.add_argument("--config", default=None, choices=["c0", "c1", "c2", "c3", "c4"],
                     help="per-configuration Lloyd iteration timing (median of iterations 2..iters)")
     ap.add_argument("--iters", type=int, default=10)
+    ap.add_argument("--hier", action="store_true",
+                    help="with --config: flat Lloyd fit against hierarchical k-means (m = sqrt k)")
     args = ap.parse_args()
     if args.case:
         run_case(args)
