@@ -85,6 +85,7 @@ def lib():
                 "or_sumsq_blocked": ([vp, i32], f64),
                 "or_split_empty_f32": ([vp, vp, i32, i32], i32),
                 "or_hadamard_rotate": ([vp, i64, i32, vp, vp, i32, vp], None),
+                "or_unproject": ([vp, i64, i32, vp, vp, i32, vp], None),
                 "or_split_empty_sq8": ([vp, vp, i32, i32], i32),
             }
             for name, (args, res) in sig.items():
@@ -338,6 +339,17 @@ def project(X, P, mu=None):
     Y = np.empty((n, dout), np.float64)
     lib().or_project(_p(X), n, d, _p(_c(mu, np.float32)) if mu is not None else None, _p(P), dout, _p(Y))
     return Y
+
+
+def unproject(Y, P, mu=None):
+    """x = y P^T + mu in fp64 (P: d x dout), [n, d]."""
+    Y = _c(Y, np.float32)
+    P = _c(P, np.float32)
+    n, dout = Y.shape
+    d = P.shape[0]
+    X = np.empty((n, d), np.float64)
+    lib().or_unproject(_p(Y), n, dout, _p(P), _p(_c(mu, np.float32)) if mu is not None else None, d, _p(X))
+    return X
 
 
 def mean_cov(X):

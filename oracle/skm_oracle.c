@@ -651,3 +651,18 @@ void or_hadamard_rotate(const float *X, int64_t n, int d, const float *mean, con
         free(v);
     }
 }
+
+/* Unprojection of projected centroids back to the original space (Section 4,
+ * "Dimensionality Reduction and Vector Search", approach 2): x = y P^T + mu,
+ * fp64, with P the d x dout projection matrix (row-major). */
+void or_unproject(const float *Y, int64_t n, int dout, const float *P, const float *mu, int d, double *X) {
+#pragma omp parallel for schedule(static)
+    for (int64_t p = 0; p < n; ++p) {
+        const float *y = Y + p * (int64_t)dout;
+        for (int i = 0; i < d; ++i) {
+            double s = mu ? (double)mu[i] : 0.0;
+            for (int j = 0; j < dout; ++j) s += (double)y[j] * (double)P[(int64_t)i * dout + j];
+            X[p * (int64_t)d + i] = s;
+        }
+    }
+}

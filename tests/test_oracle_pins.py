@@ -511,3 +511,22 @@ def test_hierarchical_recovers_separated_blobs_and_refine_does_not_hurt():
     w = oracle.objective_f32(X, C, a)
     C2, a2, _, _ = oracle.hierarchical("f32", X, 12, 4, meso_init, 3, 5, refine=True)
     assert oracle.objective_f32(X, C2, a2) <= w * (1 + 1e-9)
+
+
+def test_unproject_inverts_a_full_rank_orthogonal_projection():
+    """With an orthogonal d x d matrix, unprojecting the projection gives the
+    points back; with the top-d' PCA axes of data that lives in d' dimensions
+    it gives them back too."""
+    r = _rng(41)
+    Q, _ = np.linalg.qr(r.standard_normal((12, 12)))
+    Q = Q.astype(np.float32)
+    X = r.standard_normal((30, 12)).astype(np.float32)
+    mu = X.mean(0).astype(np.float32)
+    Y = oracle.project(X, Q, mu).astype(np.float32)
+    np.testing.assert_allclose(oracle.unproject(Y, Q, mu), X, atol=1e-5)
+    # rank-3 data in 8 dims: 3 axes suffice
+    B = np.linalg.qr(r.standard_normal((8, 3)))[0].astype(np.float32)
+    Z = (r.standard_normal((40, 3)) @ B.T + 2.0).astype(np.float32)
+    mz = Z.mean(0).astype(np.float32)
+    Yz = oracle.project(Z, B, mz).astype(np.float32)
+    np.testing.assert_allclose(oracle.unproject(Yz, B, mz), Z, atol=1e-5)
