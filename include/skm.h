@@ -128,6 +128,18 @@ size_t skm_workspace_size(int op, const skm_data *x, int k);
 int skm_project(const float *X, int64_t n, int d, const float *mean, const float *P,
                 int d_out, int out_dtype, void *Y, void *stream);
 
+/* Unprojection of centroids found in a projected space back to the original
+ * space (Section 4, "Dimensionality Reduction and Vector Search", approach 2):
+ * X = Y P^T + mean, Y float32 [n][d_out], P the projection matrix of
+ * skm_project (float32 [d][d_out], row-major), mean float32[d] or NULL, X
+ * float32 [n][d] (all device).  fp32 arithmetic; n <= 1,048,560 (centroids).
+ * Approach 1 (full-dimensional centroids from the cluster membership) and the
+ * raw-vector last update of RabitQ (Section 4, "Closing RabitQ's Gap in
+ * Balance") are skm_update on the raw float32 points with the assignment.
+ * Asynchronous. */
+int skm_unproject(const float *Y, int64_t n, int d_out, const float *P, const float *mean, int d,
+                  float *X, void *stream);
+
 /* Randomized Hadamard rotation (a structured random orthogonal transform in
  * place of a dense random rotation before RabitQ / SuperKMeans, Section 3.1;
  * O(D log D) per point): Y = (1/sqrt(D)) H_D diag(sigma) [X - mean; 0] with

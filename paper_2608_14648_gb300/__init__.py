@@ -35,7 +35,7 @@ _lib = None
 # Every entry point declared in include/skm.h.
 EXPORTED_SYMBOLS = [
     "skm_last_error", "skm_version", "skm_kernel_launches", "skm_workspace_size", "skm_screen_bytes",
-    "skm_screen_prep", "skm_project", "skm_project_hadamard", "skm_make_rotation",
+    "skm_screen_prep", "skm_project", "skm_project_hadamard", "skm_unproject", "skm_make_rotation",
     "skm_pca_fit", "skm_quantize", "skm_rbq1_exponent", "skm_assign", "skm_assign_rbq1_noalloc",
     "skm_assign_segmented",
     "skm_update",
@@ -107,6 +107,7 @@ def lib():
             "skm_project": ([vp, i64, i32, vp, vp, i32, i32, vp, vp], i32),
             "skm_make_rotation": ([u64, i32, vp], i32),
             "skm_project_hadamard": ([vp, i64, i32, vp, vp, i32, i32, vp, vp], i32),
+            "skm_unproject": ([vp, i64, i32, vp, vp, i32, vp, vp], i32),
             "skm_pca_fit": ([vp, i64, i32, i32, vp, vp, vp, vp, sz, vp], i32),
             "skm_quantize": ([i32, vp, i64, i32, vp, vp, vp, sz, vp], i32),
             "skm_rbq1_exponent": ([vp, i64, vp, vp, sz, vp], i32),
@@ -219,6 +220,15 @@ def skm_project_hadamard(X, sigma, mean=None, out_dtype=DTYPE_F32, stream=None):
     _check(lib().skm_project_hadamard(_ptr(X), n, d, _ptr(mean), _ptr(sigma), int(D), out_dtype, _ptr(Y),
                                       _stream(stream)))
     return Y
+
+
+def skm_unproject(Y, P, mean=None, stream=None):
+    """X = Y P^T + mean (P: the d x d_out projection matrix)."""
+    n, d_out = Y.shape
+    d = P.shape[0]
+    X = torch.empty(n, d, device=Y.device, dtype=torch.float32)
+    _check(lib().skm_unproject(_ptr(Y), n, d_out, _ptr(P), _ptr(mean), d, _ptr(X), _stream(stream)))
+    return X
 
 
 def skm_make_rotation(seed, d):

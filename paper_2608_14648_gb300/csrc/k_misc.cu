@@ -443,3 +443,55 @@ cudaError_t launch_hadamard(const float *X, int64_t n, int d, const float *mean,
 }
 
 }  // namespace skm
+
+namespace skm {
+
+// x = y P^T + mu (unprojection of projected centroids, Section 4 "Dimensionality
+// Reduction and Vector Search"): 16 x 64 output tiles, y rows and P rows staged
+// through shared memory in 32-wide slices; fp32 FMA.
+__global__ void __launch_bounds__(256) unproject_kernel(const float *__restrict__ Y, int64_t n, int dout,
+                                                        const float *__restrict__ P, const float *__restrict__ mu,
+                                                        int d, float *__restrict__ X) {
+    __shared__ float ys[16][33];
+    __shared__ float ps[64][33];
+    const int tx = threadIdx.x & 63, ty = threadIdx.x >> 6;  // 64 x 4 threads, 4 rows each
+    const int64_t r0 = (int64_t)blockIdx.y * 16;
+    const int c0 = blockIdx.x * 64;
+    float acc[4] = {0.f, 0.f, 0.f, 0.f};
+    for (int j0 = 0; j0 < dout; j0 += 32) {
+        __syncthreads();
+        for (int t = threadIdx.x; t < 16 * 32; t += 256) {
+            const int rr = t >> 5, jj = t & 31;
+            ys[rr][jj] = (r0 + rr < n && j0 + jj < dout) ? Y[(r0 + rr) * dout + j0 + jj] : 0.f;
+        }
+        for (int t = threadIdx.x; t < 64 * 32; t += 256) {
+            const int cc = t >> 5, jj = t & 31;
+            ps[cc][jj] = (c0 + cc < d && j0 + jj < dout) ? P[(int64_t)(c0 + cc) * dout + j0 + jj] : 0.f;
+        }
+        __syncthreads();
+#pragma unroll 8
+        for (int jj = 0; jj < 32; ++jj) {
+            const float pv = ps[tx][jj];
+#pragma unroll
+            for (int q = 0; q < 4; ++q) acc[q] = __fmaf_rn(ys[ty * 4 + q][jj], pv, acc[q]);
+        }
+    }
+    const int c = c0 + tx;
+    if (c < d)
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+            const int64_t r = r0 + ty * 4 + q;
+            if (r < n) X[r * d + c] = __fadd_rn(acc[q], mu ? mu[c] : 0.f);
+        }
+}
+
+cudaError_t launch_unproject(const float *Y, int64_t n, int dout, const float *P, const float *mu, int d,
+                             float *X, cudaStream_t st) {
+    if (n == 0) return cudaSuccess;
+    const dim3 grid((unsigned)((d + 63) / 64), (unsigned)((n + 15) / 16));
+    if (grid.y > 65535u) return cudaErrorInvalidValue;
+    unproject_kernel<<<grid, 256, 0, st>>>(Y, n, dout, P, mu, d, X);
+    return launched();
+}
+
+}  // namespace skm

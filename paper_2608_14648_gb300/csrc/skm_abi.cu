@@ -375,6 +375,15 @@ int skm_project_hadamard(const float *X, int64_t n, int d, const float *mean, co
     return SKM_OK;
 }
 
+int skm_unproject(const float *Y, int64_t n, int d_out, const float *P, const float *mean, int d, float *X,
+                  void *stream) {
+    if (!Y || !P || !X) return set_error(SKM_ERR_INVALID_ARG, "NULL pointer");
+    if (n < 1 || n > 65535LL * 16 || d < 1 || d > MAX_D || d_out < 1 || d_out > MAX_D)
+        return set_error(SKM_ERR_INVALID_ARG, "bad shape n=%lld d=%d d_out=%d", (long long)n, d, d_out);
+    SKM_CUDA_TRY(launch_unproject(Y, n, d_out, P, mean, d, X, S(stream)));
+    return SKM_OK;
+}
+
 int skm_make_rotation(uint64_t seed, int d, float *P_host) {
     if (!P_host || d < 1 || d > MAX_D) return set_error(SKM_ERR_INVALID_ARG, "bad arguments");
     std::vector<double> A((size_t)d * d);

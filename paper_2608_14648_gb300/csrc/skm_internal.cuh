@@ -166,6 +166,9 @@ cudaError_t launch_gather_rows_bytes(const void *src, int64_t rowbytes, const in
                                      void *dst, cudaStream_t st);
 // out[perm[q]] = in[q] for 4-byte values
 cudaError_t launch_unpermute(const void *in, const int32_t *perm, int64_t n, void *out, cudaStream_t st);
+// x = y P^T + mu (n <= 65535 * 16 rows)
+cudaError_t launch_unproject(const float *Y, int64_t n, int dout, const float *P, const float *mu, int d,
+                             float *X, cudaStream_t st);
 // empty clusters take half of the largest one (w: k int64 of workspace)
 cudaError_t launch_split_empty(void *C, int code_bytes, const int64_t *counts, int k, int d,
                                int64_t *w, cudaStream_t st);

@@ -676,3 +676,48 @@ def test_fit_hierarchical_f32_vs_oracle(skm):
     wg = oracle.objective_f32(X.numpy(), C.cpu().numpy(), a.cpu().numpy())
     wo = oracle.objective_f32(X.numpy(), Co, ao)
     assert abs(wg - wo) / wo <= 1e-3
+
+
+# ------------------------------------- centroids back in the original space
+@pytest.mark.parametrize("k,d,dout", [(300, 96, 32), (1000, 1024, 256), (17, 50, 50)])
+def test_unproject_vs_oracle(skm, k, d, dout):
+    g = torch.Generator().manual_seed(k + d)
+    Y = torch.randn(k, dout, generator=g)
+    P = torch.randn(d, dout, generator=g)
+    mu = torch.randn(d, generator=g)
+    X = skm.skm_unproject(Y.to(DEV), P.to(DEV), mu.to(DEV)).cpu().numpy()
+    Xo = oracle.unproject(Y.numpy(), P.numpy(), mu.numpy())
+    err = np.linalg.norm(X - Xo, axis=1) / np.maximum(np.linalg.norm(Xo, axis=1), 1e-30)
+    assert err.max() <= 1e-5
+
+
+def test_raw_vector_last_update_and_full_dimensional_centroids(skm):
+    """RabitQ's raw-vector last update and PCA's approach 1 are an update with
+    the raw float32 points and the quantized / projected run's assignment:
+    the oracle's mean of members, and (for fixed assignments) no other
+    centroids have a lower WCSS."""
+    n, d, k = 6000, 128, 40
+    X = _points(n, d, seed=61)
+    r = skm.skm_quantize(skm.REPR_RBQ1, X.to(DEV))
+    pts = skm.rbq1_points(r, d)
+    idx = synth.forgy_indices(n, k, seed=61)
+    C, a, _, _, _ = skm.skm_fit(pts, k, 4, init_idx=idx.to(DEV))
+    Craw, counts = skm.skm_update(skm.Points(skm.REPR_F32, X.to(DEV), d), a, C.clone())
+    Co, co = oracle.update_f32(X.numpy(), a.cpu().numpy(), C.cpu().numpy())
+    np.testing.assert_array_equal(counts.cpu().numpy(), co)
+    rel = np.linalg.norm(Craw.cpu().numpy() - Co, axis=1) / np.maximum(np.linalg.norm(Co, axis=1), 1e-30)
+    assert rel.max() <= 1e-4
+    ah = a.cpu().numpy()
+    assert oracle.objective_f32(X.numpy(), Craw.cpu().numpy(), ah) <= \
+        oracle.objective_f32(X.numpy(), C.cpu().numpy(), ah) * (1 + 1e-7)
+    # PCA: cluster the projection, then approach 2 (unproject) and approach 1 (members)
+    mean, P, _ = skm.skm_pca_fit(X.to(DEV), 32)
+    Yp = skm.skm_project(X.to(DEV), P, mean)
+    Cp, ap, _, _, _ = skm.skm_fit(skm.Points(skm.REPR_F32, Yp, 32), k, 4, init_idx=idx.to(DEV))
+    Cu = skm.skm_unproject(Cp, P, mean).cpu().numpy()
+    Cuo = oracle.unproject(Cp.cpu().numpy(), P.cpu().numpy(), mean.cpu().numpy())
+    np.testing.assert_allclose(Cu, Cuo, rtol=1e-5, atol=1e-6)
+    Cm, _ = skm.skm_update(skm.Points(skm.REPR_F32, X.to(DEV), d), ap, torch.from_numpy(Cu).to(DEV))
+    Cmo, _ = oracle.update_f32(X.numpy(), ap.cpu().numpy(), Cu)
+    rel = np.linalg.norm(Cm.cpu().numpy() - Cmo, axis=1) / np.maximum(np.linalg.norm(Cmo, axis=1), 1e-30)
+    assert rel.max() <= 1e-4
