@@ -87,6 +87,10 @@ def lib():
                 "or_hadamard_rotate": ([vp, i64, i32, vp, vp, i32, vp], None),
                 "or_unproject": ([vp, i64, i32, vp, vp, i32, vp], None),
                 "or_split_empty_sq8": ([vp, vp, i32, i32], i32),
+                "or_lvq4_encode": ([vp, i64, i32, vp, vp, vp], None),
+                "or_lvq4_assign": ([vp, vp, i64, i32, vp, vp, vp, i32, vp, vp], None),
+                "or_lvq4_exponent": ([vp, i64], i32),
+                "or_lvq4_update": ([vp, vp, i64, i32, i32, vp, i32, vp, vp], None),
             }
             for name, (args, res) in sig.items():
                 fn = getattr(L, name)
@@ -328,6 +332,82 @@ def rbq1_decode_points(codes, F, d, m, e, idx):
 
 
 # --------------------------------------------------------------------------
+# LVQ4 (Section 3.1 "LVQ4", Eq. final:lvq, fused decode-average)
+# --------------------------------------------------------------------------
+def lvq4_encode(V):
+    """Per-vector LVQ4 of V [n, d]: (codes uint8[n, d] in 0..15,
+    fac f32[n, 4] = (s, b, N, A), G f32[n] = s * sum(codes))."""
+    V = _c(V, np.float32)
+    n, d = V.shape
+    codes = np.empty((n, d), np.uint8)
+    fac = np.empty((n, 4), np.float32)
+    G = np.empty(n, np.float32)
+    lib().or_lvq4_encode(_p(V), n, d, _p(codes), _p(fac), _p(G))
+    return codes, fac, G
+
+
+def lvq4_pack(codes):
+    """Nibble-packed layout of 4-bit codes: uint32 [n, ceil(d/8)], dimension
+    8w + j in bits 4j .. 4j + 3 of word w, unused nibbles 0."""
+    codes = np.asarray(codes, np.uint8)
+    n, d = codes.shape
+    W = (d + 7) // 8
+    pad = np.zeros((n, 8 * W), np.uint32)
+    pad[:, :d] = codes
+    out = np.zeros((n, W), np.uint32)
+    for j in range(8):
+        out |= pad[:, j::8] << np.uint32(4 * j)
+    return out
+
+
+def lvq4_unpack(words, d):
+    words = np.asarray(words).view(np.uint32)
+    n, W = words.shape
+    out = np.empty((n, 8 * W), np.uint8)
+    for j in range(8):
+        out[:, j::8] = (words >> np.uint32(4 * j)) & np.uint32(15)
+    return out[:, :d]
+
+
+def lvq4_assign(codes, fac, prep):
+    """prep = lvq4_encode(C).  Returns (assign int32[n], dist f32[n])."""
+    codes = _c(codes, np.uint8)
+    n, d = codes.shape
+    yc, yfac, Gy = prep
+    k = yc.shape[0]
+    a = np.empty(n, np.int32)
+    dist = np.empty(n, np.float32)
+    lib().or_lvq4_assign(_p(codes), _p(_c(fac, np.float32)), n, d, _p(_c(yc, np.uint8)),
+                         _p(_c(yfac, np.float32)), _p(_c(Gy, np.float32)), k, _p(a), _p(dist))
+    return a, dist
+
+
+def lvq4_exponent(fac) -> int:
+    fac = _c(fac, np.float32)
+    return int(lib().or_lvq4_exponent(_p(fac), fac.shape[0]))
+
+
+def lvq4_update(codes, fac, e, assign, C):
+    codes = _c(codes, np.uint8)
+    n, d = codes.shape
+    Cn = np.array(C, dtype=np.float32, copy=True, order="C")
+    k = Cn.shape[0]
+    counts = np.empty(k, np.int64)
+    lib().or_lvq4_update(_p(codes), _p(_c(fac, np.float32)), n, d, int(e), _p(_c(assign, np.int32)), k,
+                         _p(Cn), _p(counts))
+    return Cn, counts
+
+
+def lvq4_decode_points(codes, fac, e, idx):
+    """Decoded points (the fused decode-average of one member each)."""
+    idx = np.asarray(idx, np.int64)
+    sub = _c(codes, np.uint8)[idx]
+    k, d = sub.shape
+    C, _ = lvq4_update(sub, _c(fac, np.float32)[idx], e, np.arange(k, dtype=np.int32), np.zeros((k, d), np.float32))
+    return C
+
+
+# --------------------------------------------------------------------------
 # Projection (rotation / PCA)
 # --------------------------------------------------------------------------
 def project(X, P, mu=None):
@@ -456,6 +536,19 @@ def lloyd_rbq1(codes, nx2, F, popx, d, m, C0, iters, e=None, split=False):
             C, _ = split_empty(C, counts)
     prep = rbq1_centroid_sq4(C, m)
     a, est = rbq1_assign(codes, nx2, F, popx, d, prep)
+    return C, a
+
+
+def lloyd_lvq4(codes, fac, C0, iters, e=None, split=False):
+    if e is None:
+        e = lvq4_exponent(fac)
+    C = np.array(C0, np.float32, copy=True)
+    for _ in range(iters):
+        a, _ = lvq4_assign(codes, fac, lvq4_encode(C))
+        C, counts = lvq4_update(codes, fac, e, a, C)
+        if split:
+            C, _ = split_empty(C, counts)
+    a, _ = lvq4_assign(codes, fac, lvq4_encode(C))
     return C, a
 
 

@@ -666,3 +666,142 @@ void or_unproject(const float *Y, int64_t n, int dout, const float *P, const flo
         }
     }
 }
+
+/* ------------------------------------------------------------------------ */
+/* Section 3.1 "LVQ4": locally-adaptive 4-bit codes with a per-vector bias   */
+/* and scale, distances by Eq. final:lvq, fused decode-average update.       */
+/* ------------------------------------------------------------------------ */
+
+/* Per vector v (a point or, once per iteration, a centroid): b = min v_i,
+ * s = (max v_i - b) / 15 in fp32 (s = 1 when the vector is flat, the same
+ * reading as the flat SQ dimension), code_i = clip(round((v_i - b) / s), 0,
+ * 15) in fp32, rounding half to even.  With S = sum code_i and
+ * Q = sum code_i^2 (exact integers) the vector's constant terms of the
+ * expanded distance are, in fp64 evaluated left to right and rounded once
+ * to fp32,
+ *   N = s*s*Q + 2*b*s*S + d*b*b     (the squared norm of the decoded vector)
+ *   A = s*S + d*b                   (the sum of the decoded vector)
+ *   G = s*S                         (s times the code sum)
+ * fac[p] = (s, b, N, A); G is returned separately (it is the centroid-side
+ * term s_y sum ybar).  Pinned: codes of data on the 15-step grid, the
+ * reconstruction error bound s/2, flat vectors, N and A against the decoded
+ * vector's fp64 norm and sum. */
+void or_lvq4_encode(const float *V, int64_t n, int d, uint8_t *codes, float *fac, float *G) {
+#pragma omp parallel for schedule(static)
+    for (int64_t p = 0; p < n; ++p) {
+        const float *v = V + p * (int64_t)d;
+        float lo = INFINITY, hi = -INFINITY;
+        for (int i = 0; i < d; ++i) {
+            if (v[i] < lo) lo = v[i];
+            if (v[i] > hi) hi = v[i];
+        }
+        float s = (hi - lo) / 15.0f;
+        if (!(s > 0.0f)) s = 1.0f;
+        int64_t S = 0, Q = 0;
+        for (int i = 0; i < d; ++i) {
+            float q = rintf((v[i] - lo) / s);
+            if (!(q >= 0.0f)) q = 0.0f;
+            if (q > 15.0f) q = 15.0f;
+            const int c = (int)q;
+            codes[p * (int64_t)d + i] = (uint8_t)c;
+            S += c;
+            Q += (int64_t)c * c;
+        }
+        const double sd = (double)s, bd = (double)lo, dd = (double)d;
+        const double N = sd * sd * (double)Q + 2.0 * bd * sd * (double)S + dd * bd * bd;
+        const double A = sd * (double)S + dd * bd;
+        fac[4 * p + 0] = s;
+        fac[4 * p + 1] = lo;
+        fac[4 * p + 2] = (float)N;
+        fac[4 * p + 3] = (float)A;
+        if (G) G[p] = (float)(sd * (double)S);
+    }
+}
+
+/* Eq. final:lvq, fp32, in this fixed order (the paper fixes none):
+ *   P   = sum_i xbar_i ybar_i                          (exact integer)
+ *   key = fma(b_y, -2 A_x, N_y)
+ *   key = fma(G_y, -2 b_x, key)                        G_y = s_y sum ybar
+ *   key = fma(-2 s_x, s_y * P, key)                    (s_y * P one rounding)
+ * The row's own N_x does not change which centroid is nearest: the argmin is
+ * taken over key (ties to the lowest index) and the reported distance is
+ * N_x + key of the winner (one fp32 addition).  xfac / yfac: (s, b, N, A)
+ * per point / centroid, Gy per centroid. */
+void or_lvq4_assign(const uint8_t *xc, const float *xfac, int64_t n, int d, const uint8_t *yc,
+                    const float *yfac, const float *Gy, int k, int32_t *assign, float *dist) {
+#pragma omp parallel for schedule(dynamic, 16)
+    for (int64_t p = 0; p < n; ++p) {
+        const uint8_t *x = xc + p * (int64_t)d;
+        const float sx2 = -2.0f * xfac[4 * p + 0];
+        const float bx2 = -2.0f * xfac[4 * p + 1];
+        const float ax2 = -2.0f * xfac[4 * p + 3];
+        float best = INFINITY;
+        int32_t a = -1;
+        for (int j = 0; j < k; ++j) {
+            const uint8_t *y = yc + (int64_t)j * d;
+            int64_t P = 0;
+            for (int i = 0; i < d; ++i) P += (int64_t)x[i] * y[i];
+            float key = fmaf(yfac[4 * j + 1], ax2, yfac[4 * j + 2]);
+            key = fmaf(Gy[j], bx2, key);
+            const float t = yfac[4 * j + 0] * (float)P;
+            key = fmaf(sx2, t, key);
+            if (key < best) {
+                best = key;
+                a = j;
+            }
+        }
+        assign[p] = a;
+        if (dist) dist[p] = xfac[4 * p + 2] + best;
+    }
+}
+
+/* Fixed-point exponent of the decode-average: with M = max over points of
+ * max(s, |b|), e = 31 - ceil(log2 M) (0 when M = 0), so that round(s 2^e) and
+ * |round(b 2^e)| are at most 2^31. */
+int or_lvq4_exponent(const float *fac, int64_t n) {
+    float mx = 0.0f;
+    for (int64_t p = 0; p < n; ++p) {
+        const float s = fac[4 * p + 0], b = fabsf(fac[4 * p + 1]);
+        if (s > mx) mx = s;
+        if (b > mx) mx = b;
+    }
+    if (!(mx > 0.0f)) return 0;
+    int ex;
+    double fr = frexp((double)mx, &ex);
+    int c = (fr == 0.5) ? ex - 1 : ex; /* ceil(log2 mx) */
+    return 31 - c;
+}
+
+/* Fused decode-average (Section 3.1 "LVQ4", last paragraph): a member decodes
+ * to s xbar_i + b and the members of a cluster are averaged.  s and b enter as
+ * the integers Sq = round(s 2^e) and Bq = round(b 2^e), so the sums are exact
+ * and independent of order:
+ *   T_i = sum Sq xbar_i,  U = sum Bq
+ *   c_i = ((T_i + U) 2^-e) / count        (int64 -> fp64, then fp32)
+ * Empty clusters keep their centroid.  Pinned against the fp64 mean of the
+ * decoded members (relative 1e-8) and exactly representable members. */
+void or_lvq4_update(const uint8_t *xc, const float *xfac, int64_t n, int d, int e,
+                    const int32_t *assign, int k, float *C_inout, int64_t *counts) {
+    int64_t *T = (int64_t *)calloc((size_t)k * d, sizeof(int64_t));
+    int64_t *U = (int64_t *)calloc((size_t)k, sizeof(int64_t));
+    for (int j = 0; j < k; ++j) counts[j] = 0;
+    for (int64_t p = 0; p < n; ++p) {
+        const int32_t a = assign[p];
+        const int64_t sq = (int64_t)llrint(ldexp((double)xfac[4 * p + 0], e));
+        const int64_t bq = (int64_t)llrint(ldexp((double)xfac[4 * p + 1], e));
+        counts[a] += 1;
+        U[a] += bq;
+        for (int i = 0; i < d; ++i) T[(int64_t)a * d + i] += sq * (int64_t)xc[p * (int64_t)d + i];
+    }
+    for (int j = 0; j < k; ++j) {
+        if (counts[j] == 0) continue;
+        for (int i = 0; i < d; ++i) {
+            double v = (double)(T[(int64_t)j * d + i] + U[j]);
+            v = ldexp(v, -e);
+            v = v / (double)counts[j];
+            C_inout[(int64_t)j * d + i] = (float)v;
+        }
+    }
+    free(T);
+    free(U);
+}

@@ -530,3 +530,169 @@ def test_unproject_inverts_a_full_rank_orthogonal_projection():
     mz = Z.mean(0).astype(np.float32)
     Yz = oracle.project(Z, B, mz).astype(np.float32)
     np.testing.assert_allclose(oracle.unproject(Yz, B, mz), Z, atol=1e-5)
+
+
+# ---------------------------------------------------------------- LVQ4
+def test_lvq4_hand_example():
+    g = json.load(open(os.path.join(GOLDEN, "lvq4_d8_hand_example.json")))
+    x = np.array([g["x"]], np.float32)
+    y = np.array([g["y"]], np.float32)
+    xc, xf, _ = oracle.lvq4_encode(x)
+    yc, yf, Gy = oracle.lvq4_encode(y)
+    assert xc[0].tolist() == g["xbar"] and yc[0].tolist() == g["ybar"]
+    assert tuple(xf[0]) == (g["s_x"], g["b_x"], g["N_x"], g["A_x"])
+    assert (yf[0, 0], yf[0, 1], yf[0, 2], Gy[0]) == (g["s_y"], g["b_y"], g["N_y"], g["G_y"])
+    assert int((xc[0].astype(np.int64) * yc[0]).sum()) == g["P"]
+    a, dist = oracle.lvq4_assign(xc, xf, (yc, yf, Gy))
+    assert a[0] == 0 and float(dist[0]) == g["distance"]
+    assert float(((x.astype(np.float64) - y) ** 2).sum()) == g["distance"]
+
+
+def _lvq4_grid(r, n, d):
+    """Vectors exactly on their own 15-step grid: power-of-two scale, bias a
+    multiple of it, codes 0 and 15 both present in every row."""
+    q = r.integers(0, 16, (n, d))
+    q[:, 0] = 0
+    q[:, 1] = 15
+    for p in range(n):
+        q[p] = q[p][r.permutation(d)]
+    s = 2.0 ** r.integers(-6, 1, n)
+    b = s * r.integers(-40, 40, n)
+    return (b[:, None] + s[:, None] * q).astype(np.float32), q, s, b
+
+
+def test_lvq4_encode_grid_exact_and_error_bound():
+    r = _rng(40)
+    X, q, s, b = _lvq4_grid(r, 50, 37)
+    codes, fac, G = oracle.lvq4_encode(X)
+    np.testing.assert_array_equal(codes, q)
+    np.testing.assert_array_equal(fac[:, 0], s.astype(np.float32))
+    np.testing.assert_array_equal(fac[:, 1], b.astype(np.float32))
+    # random vectors: codes in range, extremes at 0 and 15, error <= s/2
+    X = (r.standard_normal((200, 65)) * r.uniform(0.01, 5, (200, 1)) + r.uniform(-3, 3, (200, 1))).astype(np.float32)
+    codes, fac, G = oracle.lvq4_encode(X)
+    assert codes.max() <= 15
+    np.testing.assert_array_equal(codes[np.arange(200), X.argmin(1)], 0)
+    np.testing.assert_array_equal(codes[np.arange(200), X.argmax(1)], 15)
+    dec = fac[:, 1:2].astype(np.float64) + fac[:, 0:1].astype(np.float64) * codes
+    err = np.abs(dec - X)
+    assert np.all(err <= fac[:, 0:1] * (0.5 + 1e-5))
+    np.testing.assert_array_equal(fac[:, 1], X.min(1))
+
+
+def test_lvq4_encode_flat_vector():
+    X = np.full((2, 10), 0.75, np.float32)
+    X[1] = -3.0
+    codes, fac, G = oracle.lvq4_encode(X)
+    assert codes.max() == 0
+    np.testing.assert_array_equal(fac[:, 0], [1.0, 1.0])
+    np.testing.assert_array_equal(fac[:, 1], [0.75, -3.0])
+    np.testing.assert_array_equal(fac[:, 2], [10 * 0.75 ** 2, 90.0])
+    np.testing.assert_array_equal(fac[:, 3], [7.5, -30.0])
+    np.testing.assert_array_equal(G, [0.0, 0.0])
+
+
+def test_lvq4_terms_are_norm_and_sum_of_decoded_vector():
+    r = _rng(41)
+    X = (r.standard_normal((100, 96)) + 0.3).astype(np.float32)
+    codes, fac, G = oracle.lvq4_encode(X)
+    dec = fac[:, 1:2].astype(np.float64) + fac[:, 0:1].astype(np.float64) * codes
+    np.testing.assert_allclose(fac[:, 2], (dec ** 2).sum(1), rtol=2e-7)
+    np.testing.assert_allclose(fac[:, 3], dec.sum(1), rtol=2e-7, atol=1e-5)
+    np.testing.assert_allclose(G, fac[:, 0].astype(np.float64) * codes.sum(1), rtol=1e-7)
+
+
+def test_lvq4_distance_is_l2_of_decoded_vectors():
+    """Eq. final:lvq against the fp64 squared distance of the decoded vectors;
+    points and centroids with different scales and biases, so a swapped or
+    dropped term shows."""
+    r = _rng(42)
+    n, k, d = 300, 12, 48
+    X = (r.standard_normal((n, d)) * r.uniform(0.5, 2, (n, 1)) + r.uniform(-1, 1, (n, 1))).astype(np.float32)
+    C = (r.standard_normal((k, d)) * r.uniform(0.5, 2, (k, 1)) + r.uniform(-1, 1, (k, 1))).astype(np.float32)
+    xc, xf, _ = oracle.lvq4_encode(X)
+    prep = oracle.lvq4_encode(C)
+    yc, yf, _ = prep
+    a, dist = oracle.lvq4_assign(xc, xf, prep)
+    dx = xf[:, 1:2].astype(np.float64) + xf[:, 0:1] * xc.astype(np.float64)
+    dy = yf[:, 1:2].astype(np.float64) + yf[:, 0:1] * yc.astype(np.float64)
+    D = cdist(dx, dy, "sqeuclidean")
+    scale = xf[:, 2:3].astype(np.float64) + yf[None, :, 2]
+    true_best = D[np.arange(n), a]
+    assert np.all(np.abs(dist - true_best) <= 1e-5 * scale[np.arange(n), a] + 1e-6)
+    srt = np.sort(D, 1)
+    ok = a == D.argmin(1)
+    gap = (srt[:, 1] - srt[:, 0]) / scale.max(1)
+    assert np.all(ok | (gap < 1e-5))
+    assert ok.mean() > 0.98
+
+
+def test_lvq4_exact_grid_assignment_and_ties():
+    """Small power-of-two grids make every fp32 step exact: the argmin is the
+    brute-force one, duplicated centroids resolve to the lower index."""
+    r = _rng(43)
+    X, _, _, _ = _lvq4_grid(r, 60, 16)
+    C, _, _, _ = _lvq4_grid(r, 5, 16)
+    C = np.concatenate([C, C[2:3]])  # centroid 5 duplicates centroid 2
+    xc, xf, _ = oracle.lvq4_encode(X)
+    a, dist = oracle.lvq4_assign(xc, xf, oracle.lvq4_encode(C))
+    D = cdist(X.astype(np.float64), C.astype(np.float64), "sqeuclidean")
+    np.testing.assert_array_equal(a, D.argmin(1))
+    np.testing.assert_array_equal(dist, D.min(1).astype(np.float32))
+    assert not np.any(a == 5)
+
+
+def test_lvq4_exponent_and_update_is_mean_of_decoded_members():
+    r = _rng(44)
+    n, d, k = 400, 40, 6
+    X = (r.standard_normal((n, d)) + 0.2).astype(np.float32)
+    codes, fac, _ = oracle.lvq4_encode(X)
+    e = oracle.lvq4_exponent(fac)
+    M = float(np.maximum(fac[:, 0], np.abs(fac[:, 1])).max())
+    assert 2.0 ** 30 < M * 2.0 ** e <= 2.0 ** 31
+    a = r.integers(0, k - 1, n).astype(np.int32)  # cluster k-1 stays empty
+    C0 = r.standard_normal((k, d)).astype(np.float32)
+    C, counts = oracle.lvq4_update(codes, fac, e, a, C0)
+    dec = fac[:, 1:2].astype(np.float64) + fac[:, 0:1] * codes.astype(np.float64)
+    for j in range(k - 1):
+        np.testing.assert_allclose(C[j], dec[a == j].mean(0), rtol=1e-6, atol=1e-7)
+        assert counts[j] == (a == j).sum()
+    np.testing.assert_array_equal(C[k - 1], C0[k - 1])
+    assert counts[k - 1] == 0
+    # K = 1: the global mean of the decoded points
+    C1, _ = oracle.lvq4_update(codes, fac, e, np.zeros(n, np.int32), C0[:1])
+    np.testing.assert_allclose(C1[0], dec.mean(0), rtol=1e-6, atol=1e-7)
+    # members exactly representable in fixed point: the mean is exact
+    G, _, _, _ = _lvq4_grid(r, 4, 8)
+    gc, gf, _ = oracle.lvq4_encode(G)
+    Cg, _ = oracle.lvq4_update(gc, gf, oracle.lvq4_exponent(gf), np.zeros(4, np.int32), np.zeros((1, 8), np.float32))
+    np.testing.assert_array_equal(Cg[0], G.astype(np.float64).mean(0).astype(np.float32))
+
+
+def test_lvq4_pack_layout():
+    codes = np.zeros((2, 11), np.uint8)
+    codes[0, 0] = 1
+    codes[0, 7] = 15
+    codes[0, 8] = 3
+    codes[1, 10] = 9
+    w = oracle.lvq4_pack(codes)
+    assert w.shape == (2, 2)
+    assert int(w[0, 0]) == 1 | (15 << 28) and int(w[0, 1]) == 3
+    assert int(w[1, 1]) == 9 << 8
+    r = _rng(45)
+    c = r.integers(0, 16, (7, 29)).astype(np.uint8)
+    np.testing.assert_array_equal(oracle.lvq4_unpack(oracle.lvq4_pack(c), 29), c)
+
+
+def test_lloyd_lvq4_points_as_centroids():
+    """N = K with the decoded points as initial centroids: every point keeps
+    its own centroid (the re-encoded decoded point reproduces its codes)."""
+    r = _rng(46)
+    X = r.standard_normal((24, 32)).astype(np.float32)
+    codes, fac, _ = oracle.lvq4_encode(X)
+    e = oracle.lvq4_exponent(fac)
+    C0 = oracle.lvq4_decode_points(codes, fac, e, np.arange(24))
+    yc, _, _ = oracle.lvq4_encode(C0)
+    np.testing.assert_array_equal(yc, codes)
+    C, a = oracle.lloyd_lvq4(codes, fac, C0, 3, e=e)
+    np.testing.assert_array_equal(a, np.arange(24))
