@@ -24,7 +24,8 @@
  *    the ABI.
  *  - Distances are squared L2.  Ties in every argmin go to the LOWEST
  *    centroid index.
- *  - Limits: 1 <= d <= 4096, 1 <= k <= 65536, 1 <= n < 2^31 (RBQ1: n <= 2^24).
+ *  - Limits: 1 <= d <= 4096, 1 <= k <= 65536, 1 <= n < 2^31 (RBQ1: n <= 2^24;
+ *    LVQ4: n <= 2^26).
  */
 #ifndef SKM_H
 #define SKM_H
@@ -53,8 +54,11 @@ typedef enum skm_repr {
     SKM_REPR_SQ8 = 1,  /* uint8 SQ8 codes [n][d] (Section 3.1, per-dim b,s)  */
     SKM_REPR_RBQ1 = 2, /* RabitQ 1-bit codes uint32 [n][ceil(d/32)]
                           (bit j of word w = dimension 32w+j) + factors     */
-    SKM_REPR_BF16 = 3  /* bfloat16 bit patterns uint16 [n][d] (projected
+    SKM_REPR_BF16 = 3, /* bfloat16 bit patterns uint16 [n][d] (projected
                           points stored in bf16), fp32 centroids            */
+    SKM_REPR_LVQ4 = 4  /* LVQ 4-bit codes uint32 [n][ceil(d/8)] (dimension
+                          8w+j in bits 4j..4j+3 of word w, unused nibbles
+                          0) + per-point terms `lvq` (Section 3.1 "LVQ4")   */
 } skm_repr;
 
 typedef enum skm_dtype { SKM_DTYPE_F32 = 0, SKM_DTYPE_BF16 = 1 } skm_dtype;
@@ -81,12 +85,16 @@ typedef struct skm_data {
     const int32_t *popx;/* number of set bits            [n]                 */
     const float *m;     /* centring mean m               [d]                 */
     int32_t rbq1_exp;   /* fixed-point exponent e of the decode-average
-                           (skm_rbq1_exponent); fit() computes it itself     */
+                           (RBQ1: skm_rbq1_exponent, LVQ4: skm_lvq4_exponent);
+                           fit() computes it itself                          */
     int32_t flags;      /* SKM_FLAG_* (0 = defaults)                          */
     /* Optional screening copy for F32 / BF16 / SQ8 assignment, built once by
      * skm_screen_prep (the points never change across Lloyd iterations).
      * NULL: skm_assign builds it in its workspace on every call.            */
     const void *screen;
+    /* LVQ4 only (output of skm_quantize): per point (s, b, N, A) of
+     * Eq. final:lvq, float32 [n][4], 16-byte aligned                        */
+    const float *lvq;
 } skm_data;
 
 /* Optional per-call statistics (host struct, filled after the call's work
@@ -180,6 +188,14 @@ int skm_pca_fit(const float *X, int64_t n, int d, int d_out, float *mean, float 
  *    ||r|| / <xbar, x>; popx = set bits.  Outputs: codes uint32[n][W],
  *    W = ceil(d/32), bit j of word w = dim 32w+j (unused high bits are 0);
  *    nx2, F float[n]; popx int32[n]; m float[d].
+ *  repr = SKM_REPR_LVQ4 (Section 3.1 "LVQ4", per-vector): b = min_i x_i,
+ *    s = (max_i x_i - b) / 15 in fp32 (s = 1 for a flat vector), code_i =
+ *    clip(round((x_i - b) / s), 0, 15) in fp32, rounding half to even; with
+ *    S = sum code_i and Q = sum code_i^2 the per-point terms of Eq. final:lvq
+ *    are N = s s Q + 2 b s S + d b b and A = s S + d b, each evaluated in
+ *    fp64 left to right and rounded once to fp32.  Outputs: codes uint32
+ *    [n][ceil(d/8)] (nibbles, layout of SKM_REPR_LVQ4), lvq float [n][4] =
+ *    (s, b, N, A).  No fitted parameters (fit is ignored).
  *  X float32 [n][d].  The x rows are assumed already rotated when RabitQ's
  *  random rotation is wanted (skm_project with skm_make_rotation's P).
  * ------------------------------------------------------------------------ */
@@ -195,6 +211,7 @@ typedef struct skm_quant_params {
     float *nx2;    /* RBQ1 outputs [n]                                       */
     float *F;
     int32_t *popx;
+    float *lvq;    /* LVQ4 output [n][4] (s, b, N, A), 16-byte aligned     */
 } skm_quant_params;
 
 int skm_quantize(int repr, const float *X, int64_t n, int d, skm_quant_params *qp,
@@ -206,12 +223,21 @@ int skm_quantize(int repr, const float *X, int64_t n, int d, skm_quant_params *q
 int skm_rbq1_exponent(const float *F, int64_t n, int *e_host, void *ws, size_t ws_bytes,
                       void *stream);
 
+/* Fixed-point exponent e of the LVQ4 decode-average: with M = max over points
+ * of max(s, |b|) (lvq: float [n][4] from skm_quantize), e = 31 - ceil(log2 M)
+ * (0 when M = 0), so round(s 2^e) and |round(b 2^e)| are at most 2^31 and the
+ * per-cluster sums of up to 2^26 points are exact in int64.  Writes *e_host;
+ * synchronises. */
+int skm_lvq4_exponent(const float *lvq, int64_t n, int *e_host, void *ws, size_t ws_bytes,
+                      void *stream);
+
 /* Screening copy of the points for the tensor-core assignment (opaque
  * layout): F32 -> bf16 copy + per-point (||x~||, ||x~ - x||); SQ8 -> centred
  * codes (code - 128) in bf16 + centred squared norms; BF16 -> per-point norms
- * (plus a padded copy when d is not a multiple of 8).  skm_screen_bytes
- * returns its size (0 when the representation needs none: RBQ1, or SQ8 with
- * d > 1024); skm_screen_prep fills `screen` (device, 256-byte aligned,
+ * (plus a padded copy when d is not a multiple of 8); RBQ1 / LVQ4 (d <= 1024)
+ * -> the codes as e4m3 bytes.  skm_screen_bytes returns its size (0 when the
+ * representation needs none: SQ8, RBQ1 or LVQ4 with d > 1024);
+ * skm_screen_prep fills `screen` (device, 256-byte aligned,
  * caller-owned) from x->x.  Asynchronous. */
 size_t skm_screen_bytes(const skm_data *x);
 int skm_screen_prep(const skm_data *x, void *screen, size_t screen_bytes, void *stream);
@@ -241,6 +267,16 @@ int skm_screen_prep(const skm_data *x, void *screen, size_t screen_bytes, void *
  *          dist = fma(-2 F, u, nx2 + ny2)
  *        where P = sum_i xbar_i ybar_i is an exact integer (tensor cores in
  *        e4m3 for d <= 1024, AND + popcount beyond).
+ *   LVQ4 float [k][d] decoded centroids; per call each centroid is
+ *        re-encoded with LVQ4 exactly as skm_quantize encodes a point
+ *        (s_y, b_y, ybar, N_y; G_y = s_y sum ybar rounded once to fp32) and
+ *        Eq. final:lvq is evaluated in fp32 in the order
+ *          key = fma(b_y, -2 A_x, N_y)
+ *          key = fma(G_y, -2 b_x, key)
+ *          key = fma(-2 s_x, s_y * P, key)
+ *        with P = sum_i xbar_i ybar_i an exact integer (tensor cores in
+ *        e4m3 for d <= 1024, __dp4a beyond); the argmin is taken over key
+ *        (N_x is the same for every centroid of a row) and dist = N_x + key.
  *  assign int32[n] (required); dist float[n] (may be NULL).
  *  prev_assign int32[n] or NULL: with SKM_FLAG_PRUNE, seeds each row's
  *  pruning bound with the distance to its previous centroid (entries outside
@@ -277,8 +313,8 @@ int skm_assign_rbq1_noalloc(const skm_data *x, const float *C, int k, int32_t *a
  * of its group g = group[r] only (base: device int32[nseg + 1], base[0] = 0,
  * non-decreasing, base[nseg] <= k, every group referenced by a row non-empty),
  * with the same per-representation rules as skm_assign (F32/BF16 exact fp32
- * argmin; SQ8 and RBQ1 bit-exact), ties to the lowest index.  Tensor-core
- * paths only: SQ8 and RBQ1 need d <= 1024; no pruning flag.  Group ids
+ * argmin; SQ8, RBQ1 and LVQ4 bit-exact), ties to the lowest index.
+ * Tensor-core paths only: SQ8, RBQ1 and LVQ4 need d <= 1024; no pruning flag.  Group ids
  * outside [0, nseg) are clamped (never an out-of-bounds access); unsorted
  * groups give undefined assignments.  Workspace: skm_workspace_size(5, x, k).
  * Asynchronous. */
@@ -296,13 +332,17 @@ int skm_assign_segmented(const skm_data *x, const void *C, int k, const int32_t 
  *             / count_j) / sqrt(d) in fp64, rounded to fp32, where
  *             T_ji = sum Fq xbar_i, U_j = sum Fq, Fq = round(F 2^e) (int64,
  *             exact), e = x->rbq1_exp.
+ *   LVQ4      fused decode-average (Section 3.1 "LVQ4"): c_ji = ((T_ji +
+ *             U_j) 2^-e) / count_j in fp64, rounded to fp32, where
+ *             T_ji = sum Sq xbar_i, U_j = sum Bq, Sq = round(s 2^e),
+ *             Bq = round(b 2^e) (int64, exact), e = x->rbq1_exp.
  *  Assignments outside [0, k) are skipped (not counted, not summed).
  *  partial != NULL selects the sharded form: nothing is finalised; the
  *  cluster sums are ADDED into `partial` and the member counts into
  *  `counts` (both zeroed by the caller before the first shard) so that
  *  shards can be merged (skm_merge_partials) and finalised
  *  (skm_update_finalize).  partial layout: F32/BF16 double[k][d];
- *  SQ8 int64[k][d]; RBQ1 int64[k][d+1] (T then U).
+ *  SQ8 int64[k][d]; RBQ1 and LVQ4 int64[k][d+1] (T then U).
  * ------------------------------------------------------------------------ */
 int skm_update(const skm_data *x, const int32_t *assign, int k, void *C_inout,
                int64_t *counts, void *partial, void *ws, size_t ws_bytes, void *stream);
@@ -320,7 +360,7 @@ int skm_update_finalize(const skm_data *x, const void *partial, const int64_t *c
  * STEP 2 once more for the final assignment.
  *  cfg->iters >= 0.  Initial centroids: C_init (device, per-repr layout of
  *  skm_assign) when non-NULL, else the points init_idx[0..k) (device int64,
- *  Forgy, STEP 1): F32/BF16 rows, SQ8 codes, RBQ1 decoded points (the
+ *  Forgy, STEP 1): F32/BF16 rows, SQ8 codes, RBQ1 / LVQ4 decoded points (the
  *  decode-average of one member).
  *  An init_idx entry outside [0, n) makes the call fail with
  *  SKM_ERR_DEVICE_CHECK before any iteration; a tensor-core pipeline wait
@@ -363,8 +403,8 @@ int skm_fit(const skm_fit_config *cfg, const skm_data *x, const void *C_init,
  * final such assignment.  refine != 0 adds the optional vanilla iteration
  * over all points and all k centroids, then a final vanilla assignment.
  * Fine centroids of meso cluster i are rows sum_{j<i} k_j .. + k_i - 1.
- *  Representations: F32, SQ8 and RBQ1 (SQ8 / RBQ1 with d <= 1024); no
- *  pruning flag.  m <= min(k, 12288); k <= n.
+ *  Representations: F32, SQ8, RBQ1 and LVQ4 (SQ8 / RBQ1 / LVQ4 with
+ *  d <= 1024); no pruning flag.  m <= min(k, 12288); k <= n.
  *  Outputs (device): C_out (k rows, per-repr layout of skm_assign),
  *  assign_out int32[n]; optional meso_assign_out int32[n] (device) and
  *  fine_counts_host int32[m] (host); stats_host may be NULL.
@@ -391,7 +431,7 @@ int skm_fit_hierarchical(const skm_hier_config *cfg, const skm_data *x, const in
  * index; nothing more happens once L has fewer than 2 members): both become
  * L's centroid moved by a relative step of 2^-10 in opposite directions,
  * +eps on even and -eps on odd dimensions for j (the reverse for L), one
- * rounded fp32 multiply per element (F32/BF16/RBQ1 centroids float32[k][d]);
+ * rounded fp32 multiply per element (F32/BF16/RBQ1/LVQ4 centroids float32[k][d]);
  * SQ8 code centroids move by one code step instead (clipped to [0, 255]).
  * L then counts as ceil(n_L / 2) members and j as floor(n_L / 2) for later
  * choices; `counts` (device int64[k], from skm_update) is not modified.

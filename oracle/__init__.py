@@ -587,8 +587,9 @@ def fine_init_positions(n_i, k_i):
 
 
 def hierarchical(kind, data, k, m, meso_init, meso_iters, fine_iters, refine=False):
-    """kind 'f32' (data = X), 'sq8' (data = codes) or 'rbq1' (data = dict of
-    codes, nx2, F, popx, d, m, e).  Returns (centroids [k], assignments [n],
+    """kind 'f32' (data = X), 'sq8' (data = codes), 'rbq1' (data = dict of
+    codes, nx2, F, popx, d, m, e) or 'lvq4' (data = dict of codes (one byte per
+    dimension), fac, e).  Returns (centroids [k], assignments [n],
     meso assignments [n], fine counts per meso cluster)."""
     if kind == "f32":
         X = _c(data, np.float32)
@@ -598,6 +599,11 @@ def hierarchical(kind, data, k, m, meso_init, meso_iters, fine_iters, refine=Fal
         X = _c(data, np.uint8)
         n = X.shape[0]
         Cm, am = lloyd_sq8(X, X[meso_init], meso_iters)
+    elif kind == "lvq4":
+        r = data
+        n = r["codes"].shape[0]
+        C0 = lvq4_decode_points(r["codes"], r["fac"], r["e"], meso_init)
+        Cm, am = lloyd_lvq4(r["codes"], r["fac"], C0, meso_iters, r["e"])
     else:
         r = data
         n = r["codes"].shape[0]
@@ -618,6 +624,9 @@ def hierarchical(kind, data, k, m, meso_init, meso_iters, fine_iters, refine=Fal
             Ci, ai, _ = lloyd_f32(X[members], X[init], fine_iters)
         elif kind == "sq8":
             Ci, ai = lloyd_sq8(X[members], X[init], fine_iters)
+        elif kind == "lvq4":
+            C0 = lvq4_decode_points(r["codes"], r["fac"], r["e"], init)
+            Ci, ai = lloyd_lvq4(r["codes"][members], r["fac"][members], C0, fine_iters, r["e"])
         else:
             C0 = rbq1_decode_points(r["codes"], r["F"], r["d"], r["m"], r["e"], init)
             Ci, ai = lloyd_rbq1(r["codes"][members], r["nx2"][members], r["F"][members], r["popx"][members],
@@ -630,6 +639,8 @@ def hierarchical(kind, data, k, m, meso_init, meso_iters, fine_iters, refine=Fal
             C, a, _ = lloyd_f32(X, C, 1)
         elif kind == "sq8":
             C, a = lloyd_sq8(X, C, 1)
+        elif kind == "lvq4":
+            C, a = lloyd_lvq4(r["codes"], r["fac"], C, 1, r["e"])
         else:
             C, a = lloyd_rbq1(r["codes"], r["nx2"], r["F"], r["popx"], r["d"], r["m"], C, 1, r["e"])
     return C, a, am, kf

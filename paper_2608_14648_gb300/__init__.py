@@ -14,15 +14,15 @@ import os
 import torch
 
 __all__ = [
-    "REPR_F32", "REPR_SQ8", "REPR_RBQ1", "REPR_BF16", "SkmError", "lib", "lib_path", "Data",
+    "REPR_F32", "REPR_SQ8", "REPR_RBQ1", "REPR_BF16", "REPR_LVQ4", "SkmError", "lib", "lib_path", "Data",
     "skm_version", "skm_kernel_launches", "skm_workspace_size", "skm_project", "skm_project_hadamard",
     "skm_make_rotation", "skm_pca_fit",
-    "skm_quantize", "skm_rbq1_exponent", "skm_assign", "skm_update", "skm_merge_partials",
+    "skm_quantize", "skm_rbq1_exponent", "skm_lvq4_exponent", "skm_assign", "skm_update", "skm_merge_partials",
     "skm_update_finalize", "skm_fit", "skm_split_empty", "skm_objective", "skm_sq8_decode", "EXPORTED_SYMBOLS",
     "EMPTY_KEEP", "EMPTY_SPLIT",
 ]
 
-REPR_F32, REPR_SQ8, REPR_RBQ1, REPR_BF16 = 0, 1, 2, 3
+REPR_F32, REPR_SQ8, REPR_RBQ1, REPR_BF16, REPR_LVQ4 = 0, 1, 2, 3, 4
 FLAG_PRUNE = 1
 DTYPE_F32, DTYPE_BF16 = 0, 1
 EMPTY_KEEP, EMPTY_SPLIT = 0, 1
@@ -36,7 +36,7 @@ _lib = None
 EXPORTED_SYMBOLS = [
     "skm_last_error", "skm_version", "skm_kernel_launches", "skm_workspace_size", "skm_screen_bytes",
     "skm_screen_prep", "skm_project", "skm_project_hadamard", "skm_unproject", "skm_make_rotation",
-    "skm_pca_fit", "skm_quantize", "skm_rbq1_exponent", "skm_assign", "skm_assign_rbq1_noalloc",
+    "skm_pca_fit", "skm_quantize", "skm_rbq1_exponent", "skm_lvq4_exponent", "skm_assign", "skm_assign_rbq1_noalloc",
     "skm_assign_segmented",
     "skm_update",
     "skm_merge_partials", "skm_update_finalize", "skm_fit", "skm_split_empty", "skm_hier_workspace_size",
@@ -57,7 +57,7 @@ class Data(ctypes.Structure):
         ("repr", ctypes.c_int32), ("d", ctypes.c_int32), ("n", ctypes.c_int64),
         ("x", ctypes.c_void_p), ("nx2", ctypes.c_void_p), ("F", ctypes.c_void_p),
         ("popx", ctypes.c_void_p), ("m", ctypes.c_void_p), ("rbq1_exp", ctypes.c_int32),
-        ("flags", ctypes.c_int32), ("screen", ctypes.c_void_p),
+        ("flags", ctypes.c_int32), ("screen", ctypes.c_void_p), ("lvq", ctypes.c_void_p),
     ]
 
 
@@ -65,7 +65,7 @@ class QuantParams(ctypes.Structure):
     _fields_ = [
         ("fit", ctypes.c_int32), ("bits", ctypes.c_int32), ("b", ctypes.c_void_p),
         ("s", ctypes.c_void_p), ("m", ctypes.c_void_p), ("nx2", ctypes.c_void_p),
-        ("F", ctypes.c_void_p), ("popx", ctypes.c_void_p),
+        ("F", ctypes.c_void_p), ("popx", ctypes.c_void_p), ("lvq", ctypes.c_void_p),
     ]
 
 
@@ -111,6 +111,7 @@ def lib():
             "skm_pca_fit": ([vp, i64, i32, i32, vp, vp, vp, vp, sz, vp], i32),
             "skm_quantize": ([i32, vp, i64, i32, vp, vp, vp, sz, vp], i32),
             "skm_rbq1_exponent": ([vp, i64, vp, vp, sz, vp], i32),
+            "skm_lvq4_exponent": ([vp, i64, vp, vp, sz, vp], i32),
             "skm_assign": ([vp, vp, i32, vp, vp, vp, vp, sz, vp], i32),
             "skm_assign_rbq1_noalloc": ([vp, vp, i32, vp, vp, vp], i32),
             "skm_assign_segmented": ([vp, vp, i32, vp, vp, i32, vp, vp, vp, sz, vp], i32),
@@ -159,20 +160,22 @@ def _dev(t):
 class Points:
     """Keeps the tensors of one skm_data alive; `.ref` is the ctypes struct."""
 
-    def __init__(self, repr_, x, d, nx2=None, F=None, popx=None, m=None, rbq1_exp=0, screen=None, flags=0):
+    def __init__(self, repr_, x, d, nx2=None, F=None, popx=None, m=None, rbq1_exp=0, screen=None, flags=0,
+                 lvq=None):
         assert x.is_contiguous()
         self.repr, self.x, self.d = repr_, x, int(d)
         self.nx2, self.F, self.popx, self.m = nx2, F, popx, m
+        self.lvq = lvq
         self.n = x.shape[0]
         self.rbq1_exp = int(rbq1_exp)
         self.screen = screen
         self.flags = int(flags)
         self.ref = Data(repr_, self.d, self.n, x.data_ptr(), _ptr(nx2), _ptr(F), _ptr(popx), _ptr(m),
-                        self.rbq1_exp, self.flags, _ptr(screen))
+                        self.rbq1_exp, self.flags, _ptr(screen), _ptr(lvq))
 
     def with_flags(self, flags):
         return Points(self.repr, self.x, self.d, self.nx2, self.F, self.popx, self.m, self.rbq1_exp, self.screen,
-                      flags)
+                      flags, self.lvq)
 
     def with_screen(self, stream=None):
         """Builds the screening copy once (skm_screen_prep) and attaches it."""
@@ -182,7 +185,7 @@ class Points:
         buf = _ws(nbytes, self.device)
         _check(lib().skm_screen_prep(ctypes.byref(self.ref), _ptr(buf), buf.numel(), _stream(stream)))
         return Points(self.repr, self.x, self.d, self.nx2, self.F, self.popx, self.m, self.rbq1_exp, buf,
-                      self.flags)
+                      self.flags, self.lvq)
 
     @property
     def device(self):
@@ -264,7 +267,7 @@ def skm_quantize(repr_, X, fit=True, b=None, s=None, m=None, stream=None, out=No
         s = s if s is not None else torch.empty(d, device=dev, dtype=torch.float32)
         codes = out.get("codes")
         codes = codes if codes is not None else torch.empty(n, d, device=dev, dtype=torch.uint8)
-        qp = QuantParams(int(fit), int(bits), b.data_ptr(), s.data_ptr(), None, None, None, None)
+        qp = QuantParams(int(fit), int(bits), b.data_ptr(), s.data_ptr(), None, None, None, None, None)
         _check(lib().skm_quantize(repr_, _ptr(X), n, d, ctypes.byref(qp), _ptr(codes), _ptr(ws), ws.numel(),
                                   _stream(stream)))
         return {"codes": codes, "b": b, "s": s}
@@ -282,11 +285,38 @@ def skm_quantize(repr_, X, fit=True, b=None, s=None, m=None, stream=None, out=No
         nx2 = _o("nx2", (n,), torch.float32)
         F = _o("F", (n,), torch.float32)
         popx = _o("popx", (n,), torch.int32)
-        qp = QuantParams(int(fit), 0, None, None, m.data_ptr(), nx2.data_ptr(), F.data_ptr(), popx.data_ptr())
+        qp = QuantParams(int(fit), 0, None, None, m.data_ptr(), nx2.data_ptr(), F.data_ptr(), popx.data_ptr(), None)
         _check(lib().skm_quantize(repr_, _ptr(X), n, d, ctypes.byref(qp), _ptr(codes), _ptr(ws), ws.numel(),
                                   _stream(stream)))
         return {"codes": codes, "m": m, "nx2": nx2, "F": F, "popx": popx}
-    raise ValueError("repr must be REPR_SQ8 or REPR_RBQ1")
+    if repr_ == REPR_LVQ4:
+        W = (d + 7) // 8
+        codes = out.get("codes")
+        codes = codes if codes is not None else torch.empty(n, W, device=dev, dtype=torch.int32)
+        lvq = out.get("lvq")
+        lvq = lvq if lvq is not None else torch.empty(n, 4, device=dev, dtype=torch.float32)
+        if tuple(codes.shape) != (n, W) or tuple(lvq.shape) != (n, 4) or not codes.is_contiguous() \
+                or not lvq.is_contiguous():
+            raise ValueError("LVQ4 outputs: codes int32 [n, ceil(d/8)], lvq float32 [n, 4], contiguous")
+        qp = QuantParams(0, 0, None, None, None, None, None, None, lvq.data_ptr())
+        _check(lib().skm_quantize(repr_, _ptr(X), n, d, ctypes.byref(qp), _ptr(codes), _ptr(ws), ws.numel(),
+                                  _stream(stream)))
+        return {"codes": codes, "lvq": lvq}
+    raise ValueError("repr must be REPR_SQ8, REPR_RBQ1 or REPR_LVQ4")
+
+
+def skm_lvq4_exponent(lvq, stream=None):
+    ws = _ws(1024, lvq.device)
+    e = ctypes.c_int(0)
+    _check(lib().skm_lvq4_exponent(_ptr(lvq), lvq.shape[0], ctypes.byref(e), _ptr(ws), ws.numel(), _stream(stream)))
+    return e.value
+
+
+def lvq4_points(q, d, e=None):
+    """Points for the LVQ4 representation from skm_quantize's outputs."""
+    if e is None:
+        e = skm_lvq4_exponent(q["lvq"])
+    return Points(REPR_LVQ4, q["codes"], d, rbq1_exp=e, lvq=q["lvq"])
 
 
 def skm_rbq1_exponent(F, stream=None):

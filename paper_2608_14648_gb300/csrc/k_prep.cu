@@ -17,15 +17,6 @@ namespace skm {
 // butterfly 16, 8, 4, 2, 1) with the block sums added in order.
 constexpr int CPREP_WARPS = 4;
 
-// e4m3 encodings of the integers 0..15 (sign 0, exponent bias 7, 3 mantissa
-// bits): 0 -> 0x00, 1 -> 0x38, 2 -> 0x40, 3 -> 0x44, 4 -> 0x48, ... 15 -> 0x57.
-__device__ __forceinline__ uint8_t e4m3_of_code(uint32_t y) {
-    if (y == 0) return 0;
-    const int e = 31 - __clz(y);                // floor(log2 y), 0..3
-    const uint32_t mant = (y << (3 - e)) & 7u;  // 3 bits below the leading one
-    return (uint8_t)(((uint32_t)(e + 7) << 3) | mant);
-}
-
 // planes != nullptr: SQ4 codes as four bit planes per word (AND + popcount
 // kernel); yq != nullptr: the same codes as e4m3 bytes, row stride dq (tensor
 // kernel).

@@ -458,6 +458,101 @@ __global__ void __launch_bounds__(RS_THREADS) ring_sum_sq8_kernel(
     ring_run(codes, perm, nval, L, flag, cons);
 }
 
+// ------------------------------------------------------------- LVQ4 rows
+// T[c][i] += Sq code_i (the fused decode-average of Section 3.1 "LVQ4"),
+// T[c][d] += Bq.  Lane l holds nibble words l + 32 t (t < NW), i.e. 8
+// dimensions per word, each with an int64 accumulator (Sq < 2^32, code < 16:
+// one 32 x 32 -> 64-bit multiply-add per row and dimension).
+template <int NW>
+struct Lvq4Cons {
+    const int32_t *scl;
+    const uint32_t *sqs;  // Sq in sorted order
+    const int64_t *bqs;   // Bq in sorted order
+    unsigned long long *T;
+    int d, W;
+    unsigned long long acc[8 * NW];
+    int64_t usum;
+    int cur;
+    int64_t q0;
+    int clw, cln;
+    uint32_t sqw, sqn;
+    int64_t bqw, bqn;
+    int cnt;
+    __device__ __forceinline__ void flush(int c, int lane) {
+#pragma unroll
+        for (int t = 0; t < NW; ++t)
+#pragma unroll
+            for (int j = 0; j < 8; ++j) {
+                const int col = 8 * (lane + 32 * t) + j;
+                if (col < d && acc[8 * t + j]) atomicAdd(T + (int64_t)c * (d + 1) + col, acc[8 * t + j]);
+                acc[8 * t + j] = 0ull;
+            }
+        if (lane == 0 && usum) atomicAdd(T + (int64_t)c * (d + 1) + d, (unsigned long long)usum);
+        usum = 0;
+    }
+    __device__ __forceinline__ void start(int64_t q0_, int cnt_, int lane) {
+        q0 = q0_;
+        cnt = cnt_;
+#pragma unroll
+        for (int t = 0; t < 8 * NW; ++t) acc[t] = 0ull;
+        usum = 0;
+        clw = lane < cnt ? __ldg(scl + q0 + lane) : -1;
+        cln = 32 + lane < cnt ? __ldg(scl + q0 + 32 + lane) : -1;
+        sqw = lane < cnt ? __ldg(sqs + q0 + lane) : 0u;
+        sqn = 32 + lane < cnt ? __ldg(sqs + q0 + 32 + lane) : 0u;
+        bqw = lane < cnt ? __ldg(bqs + q0 + lane) : 0;
+        bqn = 32 + lane < cnt ? __ldg(bqs + q0 + 32 + lane) : 0;
+        cur = __shfl_sync(0xffffffffu, clw, 0);
+    }
+    __device__ __forceinline__ void row(int i, const uint8_t *slot, int lane) {
+        if ((i & 31) == 0 && i > 0) {
+            clw = cln;
+            sqw = sqn;
+            bqw = bqn;
+            const int nx = i + 32 + lane;
+            cln = nx < cnt ? __ldg(scl + q0 + nx) : -1;
+            sqn = nx < cnt ? __ldg(sqs + q0 + nx) : 0u;
+            bqn = nx < cnt ? __ldg(bqs + q0 + nx) : 0;
+        }
+        const int c = __shfl_sync(0xffffffffu, clw, i & 31);
+        const uint32_t sq = __shfl_sync(0xffffffffu, sqw, i & 31);
+        const int64_t bq = __shfl_sync(0xffffffffu, bqw, i & 31);
+        if (c != cur) {
+            flush(cur, lane);
+            cur = c;
+        }
+        usum += bq;
+        const uint32_t *words = reinterpret_cast<const uint32_t *>(slot);
+#pragma unroll
+        for (int t = 0; t < NW; ++t) {
+            const int w = lane + 32 * t;
+            if (w < W) {
+                const uint32_t v = words[w];
+#pragma unroll
+                for (int j = 0; j < 8; ++j) acc[8 * t + j] += (unsigned long long)sq * ((v >> (4 * j)) & 15u);
+            }
+        }
+    }
+    __device__ __forceinline__ void finish(int lane) { flush(cur, lane); }
+};
+
+template <int NW>
+__global__ void __launch_bounds__(RS_THREADS) ring_sum_lvq4_kernel(
+    const uint32_t *__restrict__ codes, const uint32_t *__restrict__ sqs, const int64_t *__restrict__ bqs, int d,
+    const int32_t *__restrict__ perm, const int32_t *__restrict__ scl, const int64_t *__restrict__ offsets, int k,
+    unsigned long long *__restrict__ T, RingLayout L, int32_t *flag) {
+    const int64_t nval = offsets[k];
+    if ((int64_t)blockIdx.x * RS_CW * RS_ROWS >= nval) return;
+    Lvq4Cons<NW> cons;
+    cons.scl = scl;
+    cons.sqs = sqs;
+    cons.bqs = bqs;
+    cons.T = T;
+    cons.d = d;
+    cons.W = lvq4_words(d);
+    ring_run(reinterpret_cast<const uint8_t *>(codes), perm, nval, L, flag, cons);
+}
+
 bool ring_layout(uint32_t rb, RingLayout &L) {
     if (rb == 0 || rb % 16 != 0) return false;
     L.rb = (int)rb;
@@ -588,6 +683,43 @@ cudaError_t launch_ring_sum_rbq1(const uint32_t *codes, const int64_t *fqs, int6
         RS_CASE(6)
         RS_CASE(7)
         RS_CASE(8)
+    default:
+        break;
+    }
+#undef RS_CASE
+    return cudaErrorInvalidValue;
+}
+
+bool ring_sum_lvq4_ok(const void *codes, int d) {
+    RingLayout L;
+    const int W = lvq4_words(d);
+    return W % 4 == 0 && W <= 128 && (reinterpret_cast<uintptr_t>(codes) & 15u) == 0 &&
+           ring_layout((uint32_t)W * 4u, L);
+}
+
+cudaError_t launch_ring_sum_lvq4(const uint32_t *codes, const uint32_t *sq, const int64_t *bq, int64_t n, int d,
+                                 const int32_t *perm, const int32_t *scl, const int64_t *offsets, int k, int64_t *T,
+                                 int32_t *flag, cudaStream_t st) {
+    if (n == 0) return cudaSuccess;
+    const int W = lvq4_words(d);
+    RingLayout L;
+    if (!ring_layout((uint32_t)W * 4u, L)) return cudaErrorInvalidValue;
+    const size_t smem = L.bytes();
+    const unsigned g = ring_blocks(n);
+    auto T64 = reinterpret_cast<unsigned long long *>(T);
+#define RS_CASE(NWV)                                                                                \
+    case NWV: {                                                                                     \
+        auto kern = ring_sum_lvq4_kernel<NWV>;                                                      \
+        cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem); \
+        if (e != cudaSuccess) return e;                                                             \
+        kern<<<g, RS_THREADS, smem, st>>>(codes, sq, bq, d, perm, scl, offsets, k, T64, L, flag);    \
+        return launched();                                                                          \
+    }
+    switch ((W + 31) / 32) {
+        RS_CASE(1)
+        RS_CASE(2)
+        RS_CASE(3)
+        RS_CASE(4)
     default:
         break;
     }

@@ -52,14 +52,17 @@ constexpr int B_STAGE = BN * BK * 2;  // 32 KiB
 constexpr int TCAND = 4;
 constexpr unsigned long long WAIT_LIMIT_NS = 2000000000ull;  // 2 s per barrier wait
 
-enum { MODE_SCREEN = 0, MODE_SQ8 = 1, MODE_RBQ1 = 2 };
+enum { MODE_SCREEN = 0, MODE_SQ8 = 1, MODE_RBQ1 = 2, MODE_LVQ4 = 3 };
 // epilogue warps per TMEM lane quarter, and CTAs per cluster (centroid
 // slices multicast across the cluster), by mode.  Clusters of 2 run
 // correctly but measured slower on GB300 (the pair's pipelines wait on each
 // other's slowest epilogue: fp32 0.999 vs 0.956 ms, 1-bit 0.602 vs 0.554 ms
 // at 1M x 1000 x 768), so every mode runs one CTA per cluster.
-constexpr int TC_NH[3] = {4, 2, 4};
-constexpr int TC_CL[3] = {1, 1, 1};
+constexpr int TC_NH[4] = {4, 2, 4, 4};
+constexpr int TC_CL[4] = {1, 1, 1, 1};
+// the e4m3 (kind::f8f6f4) modes: 128 elements per 128-byte K slice
+template <int MODE>
+constexpr bool f8_mode() { return MODE == MODE_RBQ1 || MODE == MODE_LVQ4; }
 
 // Epilogue shape: NH warps per TMEM lane quarter (column slices of 256 / NH).
 template <int NH>
@@ -103,6 +106,8 @@ struct TcParams {
     const float *nx2;        // RBQ1 per point
     const float *F;
     const int32_t *popx;
+    const float4 *lvq;       // LVQ4 per point (s, b, N, A); rinfo / rinfoq hold
+                             // the column pairs (b x2, G x2) / (s x2, N x2)
     int d;
     // Segmented mode (all NULL otherwise): the point rows are sorted by
     // group and row r may only take centroids [seg_base[g], seg_base[g + 1])
@@ -404,7 +409,7 @@ __global__ void __launch_bounds__(tc_threads<NH>(), 1)
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     volatile int32_t *abort_flag = p.counters + 2;
-    constexpr int KC_ELEMS = (MODE == MODE_RBQ1) ? 128 : 64;  // elements per 128-byte row
+    constexpr int KC_ELEMS = f8_mode<MODE>() ? 128 : 64;  // elements per 128-byte row
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < STAGES; ++s) {
@@ -485,7 +490,7 @@ __global__ void __launch_bounds__(tc_threads<NH>(), 1)
                         const uint64_t bd = sw128_desc(sB + s * B_STAGE);
 #pragma unroll
                         for (int kk = 0; kk < 4; ++kk) {  // 4 x 32-byte K steps per 128-byte row
-                            if (MODE == MODE_RBQ1)
+                            if (f8_mode<MODE>())
                                 tc_mma_f8(dcol, ad + 2u * kk, bd + 2u * kk, IDESC_F8, (kc | kk) != 0);
                             else
                                 tc_mma(dcol, ad + 2u * kk, bd + 2u * kk, IDESC, (kc | kk) != 0);
@@ -525,7 +530,7 @@ __global__ void __launch_bounds__(tc_threads<NH>(), 1)
                     const float4 ci = __ldg(p.cinfo + ctn * 128 + te);
                     pre2 = make_float2(ci.x, ci.y);
                 }
-            } else if (MODE == MODE_RBQ1) {
+            } else if (f8_mode<MODE>()) {
                 if (te < 128) pre4 = __ldg(p.rinfo + ctn * 128 + te);
                 else if (te < 256) pre4 = __ldg(p.rinfoq + ctn * 128 + (te - 128));
             } else {
@@ -536,7 +541,7 @@ __global__ void __launch_bounds__(tc_threads<NH>(), 1)
             uint8_t *rb = rec_base + buf * REC_BYTES;
             if (MODE == MODE_SCREEN) {
                 if (te < 128) reinterpret_cast<float2 *>(rb)[te] = pre2;
-            } else if (MODE == MODE_RBQ1) {
+            } else if (f8_mode<MODE>()) {
                 if (te < 256) reinterpret_cast<float4 *>(rb)[te] = pre4;
             } else {
                 if (te < 256) reinterpret_cast<int32_t *>(rb)[te] = pre1;
@@ -582,6 +587,13 @@ __global__ void __launch_bounds__(tc_threads<NH>(), 1)
                 w2 = 2.0f * __fmaf_ru(a2, __ldg(p.hz), __ldg(p.hz + 1));
             } else if (MODE == MODE_SQ8) {
                 nxr = valid ? p.nx[row] : 0;
+            } else if (MODE == MODE_LVQ4) {
+                // per row: -2 s_x, -2 b_x, -2 A_x (exact) and N_x
+                const float4 f = valid ? p.lvq[row] : make_float4(0.f, 0.f, 0.f, 0.f);
+                rpc = __fmul_rn(-2.0f, f.x);
+                rf2 = __fmul_rn(-2.0f, f.y);
+                a2 = __fmul_rn(-2.0f, f.w);
+                rnx2 = f.z;
             } else {
                 rnx2 = valid ? p.nx2[row] : 0.0f;
                 rf2 = valid ? __fmul_rn(-2.0f, p.F[row]) : 0.0f;  // exact
@@ -672,6 +684,51 @@ __global__ void __launch_bounds__(tc_threads<NH>(), 1)
                                 besti = j0 + i;
                             }
                         }
+                    } else if (MODE == MODE_LVQ4) {
+                        // Eq. final:lvq in the library's fixed fp32 order:
+                        // key = fma(b_y, -2 A_x, N_y); key = fma(G_y, -2 b_x, key);
+                        // key = fma(-2 s_x, s_y P, key).  P is the nearest integer
+                        // to the e4m3 accumulator ((acc + 2^23) - 2^23, exact for
+                        // 0 <= acc < 2^22; P <= 225 d).  Two columns per packed op.
+                        float gb[4];
+                        int gi[4];
+#pragma unroll
+                        for (int g = 0; g < 4; ++g) {
+                            asm volatile("" ::: "memory");
+                            gb[g] = INFINITY;
+                            gi[g] = 0x7fffffff;
+#pragma unroll
+                            for (int i = 8 * g; i < 8 * g + 8; i += 2) {
+                                const float4 bg = reinterpret_cast<const float4 *>(rbuf)[(cc + i) >> 1];
+                                const float4 sn = reinterpret_cast<const float4 *>(rbuf)[128 + ((cc + i) >> 1)];
+                                const float2 P2 = fsub2(
+                                    fadd2(make_float2(__uint_as_float(v[i]), __uint_as_float(v[i + 1])),
+                                          make_float2(0x1p23f, 0x1p23f)),
+                                    make_float2(0x1p23f, 0x1p23f));
+                                float2 key = ffma2(make_float2(bg.x, bg.y), make_float2(a2, a2), make_float2(sn.z, sn.w));
+                                key = ffma2(make_float2(bg.z, bg.w), make_float2(rf2, rf2), key);
+                                const float2 t = fmul2(make_float2(sn.x, sn.y), P2);
+                                key = ffma2(make_float2(rpc, rpc), t, key);
+                                if (SEG && (j0 < cb || j0 + 32 > ce)) {  // columns outside the row's group
+                                    if (j0 + i < cb || j0 + i >= ce) key.x = INFINITY;
+                                    if (j0 + i + 1 < cb || j0 + i + 1 >= ce) key.y = INFINITY;
+                                }
+                                if (key.x < gb[g]) {
+                                    gb[g] = key.x;
+                                    gi[g] = j0 + i;
+                                }
+                                if (key.y < gb[g]) {
+                                    gb[g] = key.y;
+                                    gi[g] = j0 + i + 1;
+                                }
+                            }
+                        }
+#pragma unroll
+                        for (int g = 0; g < 4; ++g)
+                            if (gb[g] < fbest) {
+                                fbest = gb[g];
+                                besti = gi[g];
+                            }
                     } else {
                         // Eq. final:rabitq in Eq. rabitq_l2 in the library's fixed
                         // fp32 order (u = fma(sd, 2P - sum ybar, bd pc),
@@ -826,6 +883,9 @@ __global__ void __launch_bounds__(tc_threads<NH>(), 1)
                 } else if (MODE == MODE_SQ8) {
                     p.assign[row] = besti;
                     if (p.dist) p.dist[row] = (float)best;
+                } else if (MODE == MODE_LVQ4) {
+                    p.assign[row] = besti;
+                    if (p.dist) p.dist[row] = __fadd_rn(rnx2, fbest);
                 } else {
                     p.assign[row] = besti;
                     if (p.dist) p.dist[row] = fbest;
@@ -1276,7 +1336,7 @@ int launch_tc(const void *xs, int64_t n, int dp, int d, const void *cs, int k, c
     // per device: the attribute and the number of clusters that fit at once
     constexpr int MAXDEV = 64;
     static std::mutex mu;
-    static int cached_clusters[3][2][MAXDEV] = {};
+    static int cached_clusters[4][2][MAXDEV] = {};
     int dev = 0;
     SKM_CUDA_TRY(cudaGetDevice(&dev));
     int max_clusters = 0;
@@ -1306,7 +1366,7 @@ int launch_tc(const void *xs, int64_t n, int dp, int d, const void *cs, int k, c
         }
     }
     CUtensorMap ma, mb;
-    const int eb = MODE == MODE_RBQ1 ? 1 : 2;
+    const int eb = f8_mode<MODE>() ? 1 : 2;
     SKM_TRY(make_map(&ma, xs, n, d, dp, BM, eb));
     SKM_TRY(make_map(&mb, cs, k, d, dp, BN / CL, eb));
     TcParams p = p0;
@@ -1369,6 +1429,10 @@ size_t tc_screen_bytes(int repr, int64_t n, int d, const void *x) {
         if (d > TC_RBQ1_MAX_D) return 0;
         cv.take<uint8_t>((size_t)n * round16(d));
         break;
+    case SKM_REPR_LVQ4:
+        if (d > TC_LVQ4_MAX_D) return 0;
+        cv.take<uint8_t>((size_t)n * round16(d));
+        break;
     default:
         return 0;
     }
@@ -1405,6 +1469,7 @@ static ScreenView screen_view(int repr, int64_t n, int d, const void *x, const v
         v.rho_max = cv.take<float>(1);
         break;
     case SKM_REPR_RBQ1:
+    case SKM_REPR_LVQ4:
         v.xs = cv.take<uint8_t>((size_t)n * round16(d));
         break;
     }
@@ -1439,6 +1504,9 @@ int tc_screen_prep(const skm_data *x, void *screen, cudaStream_t st) {
                                                              d, round16(d), (uint8_t *)v.xs);
         break;
     }
+    case SKM_REPR_LVQ4:
+        SKM_CUDA_TRY(launch_lvq4_expand(static_cast<const uint32_t *>(x->x), n, d, (uint8_t *)v.xs, round16(d), st));
+        return SKM_OK;
     default:
         return set_error(SKM_ERR_INVALID_ARG, "no screening copy for repr %d", x->repr);
     }
@@ -1454,6 +1522,7 @@ void tc_plan(int repr, int64_t n, int d, int k, const void *x, const void *scree
     const int dp = round8(d);
     const bool dense = repr == SKM_REPR_F32 || repr == SKM_REPR_BF16 ||
                        (repr == SKM_REPR_RBQ1 && d <= TC_RBQ1_MAX_D) ||
+                       (repr == SKM_REPR_LVQ4 && d <= TC_LVQ4_MAX_D) ||
                        (repr == SKM_REPR_SQ8 && d <= TC_SQ8_MAX_D);
     if (!dense) return;
     if (!screen) {
@@ -1461,6 +1530,13 @@ void tc_plan(int repr, int64_t n, int d, int k, const void *x, const void *scree
         b.screen = cv.take<uint8_t>(sb);
     }
     const size_t kp = (size_t)cdiv(k, BN) * BN;  // per-centroid records padded to whole tiles
+    if (repr == SKM_REPR_LVQ4) {
+        b.cs = reinterpret_cast<uint16_t *>(cv.take<uint8_t>((size_t)k * round16(d)));
+        b.linfo = cv.take<float4>(k);
+        b.rpair_bs = cv.take<float4>(kp / 2);
+        b.rpair_qn = cv.take<float4>(kp / 2);
+        return;
+    }
     if (repr == SKM_REPR_RBQ1) {
         b.cs = reinterpret_cast<uint16_t *>(cv.take<uint8_t>((size_t)k * round16(d)));
         b.rinfo = cv.take<Rbq1CInfo>(k);
@@ -1642,6 +1718,35 @@ int tc_assign_rbq1(const skm_data *x, const float *C, int k, int32_t *assign, fl
     p.d = d;
     SKM_TRY(seg_setup(seg, n, p, st));
     SKM_TRY(launch_tc<MODE_RBQ1>(v.xs, n, dp, d, b.cs, k, p, st));
+    add_stats_kernel<<<1, 1, 0, st>>>(b.counters, b.stats);
+    SKM_CUDA_TRY(launched());
+    return SKM_OK;
+}
+
+int tc_assign_lvq4(const skm_data *x, const float *C, int k, int32_t *assign, float *dist,
+                   TcAssignBufs &b, cudaStream_t st, const TcSeg *seg) {
+    const int64_t n = x->n;
+    const int d = x->d, dp = round16(d);
+    const void *screen = x->screen;
+    if (!screen) {
+        SKM_TRY(tc_screen_prep(x, b.screen, st));
+        screen = b.screen;
+    }
+    ScreenView v = screen_view(x->repr, n, d, x->x, screen);
+    const int kp = (int)(cdiv(k, BN) * BN);
+    SKM_CUDA_TRY(launch_lvq4_cprep(C, k, d, reinterpret_cast<uint8_t *>(b.cs), dp, nullptr, b.linfo, st));
+    SKM_CUDA_TRY(launch_lvq4_pack_pairs(b.linfo, k, kp, b.rpair_bs, b.rpair_qn, st));
+    SKM_CUDA_TRY(cudaMemsetAsync(b.counters, 0, sizeof(int32_t) * 4, st));
+    TcParams p{};
+    p.counters = b.counters;
+    p.assign = assign;
+    p.dist = dist;
+    p.rinfo = b.rpair_bs;
+    p.rinfoq = b.rpair_qn;
+    p.lvq = reinterpret_cast<const float4 *>(x->lvq);
+    p.d = d;
+    SKM_TRY(seg_setup(seg, n, p, st));
+    SKM_TRY(launch_tc<MODE_LVQ4>(v.xs, n, dp, d, b.cs, k, p, st));
     add_stats_kernel<<<1, 1, 0, st>>>(b.counters, b.stats);
     SKM_CUDA_TRY(launched());
     return SKM_OK;

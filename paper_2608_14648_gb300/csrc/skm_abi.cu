@@ -36,12 +36,13 @@ constexpr int MAX_D = 4096;
 constexpr int MAX_K = 65536;
 constexpr int64_t MAX_N = (int64_t(1) << 31) - 1;
 constexpr int64_t MAX_N_RBQ1 = int64_t(1) << 24;
+constexpr int64_t MAX_N_LVQ4 = int64_t(1) << 26;
 constexpr int RED_BLOCKS = 304;
 constexpr int PRUNE_MAX_D = 1024;  // 2 x 152 SMs for column / objective reductions
 
 static int check_data(const skm_data *x, bool need_codes = true) {
     if (!x) return set_error(SKM_ERR_INVALID_ARG, "skm_data is NULL");
-    if (x->repr < SKM_REPR_F32 || x->repr > SKM_REPR_BF16)
+    if (x->repr < SKM_REPR_F32 || x->repr > SKM_REPR_LVQ4)
         return set_error(SKM_ERR_INVALID_ARG, "unknown repr %d", x->repr);
     if (x->d < 1 || x->d > MAX_D)
         return set_error(x->d < 1 ? SKM_ERR_INVALID_ARG : SKM_ERR_UNSUPPORTED,
@@ -59,6 +60,13 @@ static int check_data(const skm_data *x, bool need_codes = true) {
                              (long long)x->n);
         if (!x->nx2 || !x->F || !x->popx || !x->m)
             return set_error(SKM_ERR_INVALID_ARG, "RBQ1 needs nx2, F, popx and m");
+    }
+    if (x->repr == SKM_REPR_LVQ4) {
+        if (x->n > MAX_N_LVQ4)
+            return set_error(SKM_ERR_UNSUPPORTED, "LVQ4 supports n <= 2^26 (got %lld)", (long long)x->n);
+        if (!x->lvq) return set_error(SKM_ERR_INVALID_ARG, "LVQ4 needs the per-point terms lvq");
+        if (((uintptr_t)x->lvq & 15) != 0)
+            return set_error(SKM_ERR_INVALID_ARG, "LVQ4 terms lvq must be 16-byte aligned");
     }
     return SKM_OK;
 }
@@ -82,6 +90,8 @@ struct AssignBufs {
     int32_t *nx = nullptr, *nc = nullptr;  // SQ8 with d > 1024 (__dp4a path)
     uint4 *planes = nullptr;                // RBQ1 with d > 1024 (AND + popcount path)
     Rbq1CInfo *info = nullptr;
+    uint32_t *yw = nullptr;                 // LVQ4 with d > 1024 (__dp4a path): centroid nibbles
+    float4 *linfo = nullptr;
     TcAssignBufs tc;                        // tensor-core paths (F32, BF16, SQ8, RBQ1)
 };
 
@@ -106,6 +116,12 @@ static void plan_assign(const skm_data *x, int k, Carver &cv, AssignBufs &b) {
             b.info = cv.take<Rbq1CInfo>(k);
         }
         break;
+    case SKM_REPR_LVQ4:
+        if (d > TC_LVQ4_MAX_D) {
+            b.yw = cv.take<uint32_t>((size_t)k * lvq4_words(d));
+            b.linfo = cv.take<float4>(k);
+        }
+        break;
     default:
         break;
     }
@@ -116,6 +132,8 @@ struct UpdateBufs {
     int32_t *counts32 = nullptr, *cursor = nullptr, *perm = nullptr, *scl = nullptr;
     int64_t *offsets = nullptr;
     int64_t *fq = nullptr;    // RBQ1: fixed-point weights round(F 2^e)
+    uint32_t *sq = nullptr;   // LVQ4: round(s 2^e), sorted order
+    int64_t *bq = nullptr;    // LVQ4: round(b 2^e), sorted order
     float *sumf = nullptr;    // F32/BF16: cluster sums [k][d]
     int64_t *sumi = nullptr;  // RBQ1: cluster sums [k][d + 1]; SQ8: [k][d]
     int32_t *flag = nullptr;  // raised by a streamed-sum wait that gave up
@@ -130,6 +148,11 @@ static void plan_update(const skm_data *x, int k, Carver &cv, UpdateBufs &b) {
     b.scl = cv.take<int32_t>(x->n);
     if (x->repr == SKM_REPR_RBQ1) {
         b.fq = cv.take<int64_t>(x->n);
+        b.sumi = cv.take<int64_t>((size_t)k * (x->d + 1));
+    }
+    if (x->repr == SKM_REPR_LVQ4) {
+        b.sq = cv.take<uint32_t>(x->n);
+        b.bq = cv.take<int64_t>(x->n);
         b.sumi = cv.take<int64_t>((size_t)k * (x->d + 1));
     }
     if (x->repr == SKM_REPR_SQ8) b.sumi = cv.take<int64_t>((size_t)k * x->d);
@@ -213,6 +236,16 @@ static int do_assign(const skm_data *x, const void *C, int k, const int32_t *pre
                                             x->popx, n, d, b.planes, b.info, k, assign, dist, st));
         }
         break;
+    case SKM_REPR_LVQ4:
+        if (d <= TC_LVQ4_MAX_D) {
+            SKM_TRY(tc_assign_lvq4(x, static_cast<const float *>(C), k, assign, dist, b.tc, st));
+        } else {
+            SKM_CUDA_TRY(launch_lvq4_cprep(static_cast<const float *>(C), k, d, nullptr, 0, b.yw, b.linfo, st));
+            SKM_CUDA_TRY(launch_assign_lvq4_simt(static_cast<const uint32_t *>(x->x),
+                                                 reinterpret_cast<const float4 *>(x->lvq), n, d, b.yw, b.linfo, k,
+                                                 assign, dist, st));
+        }
+        break;
     }
     return SKM_OK;
 }
@@ -268,6 +301,19 @@ static int do_update(const skm_data *x, const int32_t *assign, int k, void *C, i
             SKM_CUDA_TRY(launch_chunk_sum_rbq1(codes, b.fq, n, d, b.perm, b.scl, b.offsets, k, T, st));
         if (!partial)
             SKM_CUDA_TRY(launch_finalize_rbq1(T, counts, k, d, x->m, e, static_cast<float *>(C), st));
+        break;
+    }
+    case SKM_REPR_LVQ4: {
+        SKM_CUDA_TRY(launch_lvq4_q(reinterpret_cast<const float4 *>(x->lvq), b.perm, b.offsets, k, n, e, b.sq, b.bq,
+                                   st));
+        int64_t *T = partial ? static_cast<int64_t *>(partial) : b.sumi;
+        if (!partial) SKM_CUDA_TRY(cudaMemsetAsync(T, 0, sizeof(int64_t) * (size_t)k * (d + 1), st));
+        const uint32_t *codes = static_cast<const uint32_t *>(x->x);
+        if (ring_sum_lvq4_ok(codes, d))
+            SKM_CUDA_TRY(launch_ring_sum_lvq4(codes, b.sq, b.bq, n, d, b.perm, b.scl, b.offsets, k, T, b.flag, st));
+        else
+            SKM_CUDA_TRY(launch_chunk_sum_lvq4(codes, b.sq, b.bq, n, d, b.perm, b.scl, b.offsets, k, T, st));
+        if (!partial) SKM_CUDA_TRY(launch_finalize_lvq4(T, counts, k, d, e, static_cast<float *>(C), st));
         break;
     }
     }
@@ -476,7 +522,30 @@ int skm_quantize(int repr, const float *X, int64_t n, int d, skm_quant_params *q
                                         qp->F, qp->popx, st));
         return SKM_OK;
     }
-    return set_error(SKM_ERR_INVALID_ARG, "skm_quantize: repr must be SQ8 or RBQ1");
+    if (repr == SKM_REPR_LVQ4) {
+        if (n > MAX_N_LVQ4) return set_error(SKM_ERR_UNSUPPORTED, "LVQ4 supports n <= 2^26");
+        if (!qp->lvq) return set_error(SKM_ERR_INVALID_ARG, "LVQ4 needs lvq");
+        if (((uintptr_t)qp->lvq & 15) != 0 || ((uintptr_t)codes & 3) != 0)
+            return set_error(SKM_ERR_INVALID_ARG, "LVQ4 outputs: lvq 16-byte, codes 4-byte aligned");
+        SKM_CUDA_TRY(launch_lvq4_encode(X, n, d, static_cast<uint32_t *>(codes), reinterpret_cast<float4 *>(qp->lvq),
+                                        st));
+        return SKM_OK;
+    }
+    return set_error(SKM_ERR_INVALID_ARG, "skm_quantize: repr must be SQ8, RBQ1 or LVQ4");
+}
+
+int skm_lvq4_exponent(const float *lvq, int64_t n, int *e_host, void *ws, size_t ws_bytes, void *stream) {
+    if (!lvq || !e_host || n < 1) return set_error(SKM_ERR_INVALID_ARG, "bad arguments");
+    if (((uintptr_t)lvq & 15) != 0) return set_error(SKM_ERR_INVALID_ARG, "lvq must be 16-byte aligned");
+    cudaStream_t st = S(stream);
+    Carver cv(ws, ws_bytes);
+    unsigned int *mb = cv.take<unsigned int>(1);
+    int *ed = cv.take<int>(1);
+    SKM_TRY(need_ws(cv, ws_bytes, ws));
+    SKM_CUDA_TRY(launch_lvq4_exponent(reinterpret_cast<const float4 *>(lvq), n, mb, ed, st));
+    SKM_CUDA_TRY(cudaMemcpyAsync(e_host, ed, sizeof(int), cudaMemcpyDeviceToHost, st));
+    SKM_CUDA_TRY(cudaStreamSynchronize(st));
+    return SKM_OK;
 }
 
 int skm_rbq1_exponent(const float *F, int64_t n, int *e_host, void *ws, size_t ws_bytes,
@@ -538,6 +607,10 @@ static int do_assign_seg(const skm_data *x, const void *C, int k, const int32_t 
         return tc_assign_float(x, static_cast<const float *>(C), k, assign, dist, b.tc, st, &sg);
     case SKM_REPR_SQ8:
         return tc_assign_sq8(x, static_cast<const uint8_t *>(C), k, b.nx, b.nc, assign, dist, b.tc, st, &sg);
+    case SKM_REPR_LVQ4:
+        if (x->d > TC_LVQ4_MAX_D)
+            return set_error(SKM_ERR_UNSUPPORTED, "segmented LVQ4 assignment needs d <= %d", TC_LVQ4_MAX_D);
+        return tc_assign_lvq4(x, static_cast<const float *>(C), k, assign, dist, b.tc, st, &sg);
     default:
         if (x->d > TC_RBQ1_MAX_D)
             return set_error(SKM_ERR_UNSUPPORTED, "segmented RBQ1 assignment needs d <= %d", TC_RBQ1_MAX_D);
@@ -570,6 +643,8 @@ static int64_t row_bytes(const skm_data *x) {
         return x->d;
     case SKM_REPR_RBQ1:
         return 4LL * words_of(x->d);
+    case SKM_REPR_LVQ4:
+        return 4LL * lvq4_words(x->d);
     default:
         return 2LL * x->d;
     }
@@ -584,6 +659,7 @@ struct HierBufs {
     uint8_t *rows = nullptr;  // the points in meso order
     float *nx2 = nullptr, *F = nullptr;
     int32_t *popx = nullptr;
+    float4 *lvq = nullptr;  // LVQ4 per-point terms in meso order
     uint8_t *screen = nullptr;
     AssignBufs a;
     int32_t *ct0 = nullptr, *nct = nullptr;
@@ -618,6 +694,7 @@ static void plan_hier(const skm_data *x, int k, int m, Carver &cv, HierBufs &b) 
         b.F = cv.take<float>(n);
         b.popx = cv.take<int32_t>(n);
     }
+    if (x->repr == SKM_REPR_LVQ4) b.lvq = cv.take<float4>(n);
     skm_data xs = *x;
     xs.x = b.rows;
     const size_t sb = tc_screen_bytes(x->repr, n, x->d, b.rows ? b.rows : reinterpret_cast<const void *>(16));
@@ -645,8 +722,9 @@ static int hier_check(const skm_hier_config *cfg, const skm_data *x) {
         return set_error(SKM_ERR_INVALID_ARG, "bad iteration counts");
     if (x->repr == SKM_REPR_BF16) return set_error(SKM_ERR_UNSUPPORTED, "hierarchical fit: F32, SQ8 or RBQ1 points");
     if (use_prune(x)) return set_error(SKM_ERR_UNSUPPORTED, "hierarchical fit has no pruning variant");
-    if ((x->repr == SKM_REPR_SQ8 && x->d > TC_SQ8_MAX_D) || (x->repr == SKM_REPR_RBQ1 && x->d > TC_RBQ1_MAX_D))
-        return set_error(SKM_ERR_UNSUPPORTED, "hierarchical SQ8 / RBQ1 fit needs d <= 1024");
+    if ((x->repr == SKM_REPR_SQ8 && x->d > TC_SQ8_MAX_D) || (x->repr == SKM_REPR_RBQ1 && x->d > TC_RBQ1_MAX_D) ||
+        (x->repr == SKM_REPR_LVQ4 && x->d > TC_LVQ4_MAX_D))
+        return set_error(SKM_ERR_UNSUPPORTED, "hierarchical SQ8 / RBQ1 / LVQ4 fit needs d <= 1024");
     return SKM_OK;
 }
 
@@ -739,6 +817,15 @@ int skm_fit_hierarchical(const skm_hier_config *cfg, const skm_data *x, const in
         SKM_CUDA_TRY(cudaStreamSynchronize(st));
         xs.rbq1_exp = e;
     }
+    if (x->repr == SKM_REPR_LVQ4) {
+        SKM_CUDA_TRY(launch_gather_rows_bytes(x->lvq, 16, b.perm, n, b.lvq, st));
+        xs.lvq = reinterpret_cast<const float *>(b.lvq);
+        SKM_CUDA_TRY(launch_lvq4_exponent(reinterpret_cast<const float4 *>(x->lvq), n, b.maxbits, b.e_dev, st));
+        int e = 0;
+        SKM_CUDA_TRY(cudaMemcpyAsync(&e, b.e_dev, sizeof(int), cudaMemcpyDeviceToHost, st));
+        SKM_CUDA_TRY(cudaStreamSynchronize(st));
+        xs.rbq1_exp = e;
+    }
     SKM_TRY(tc_screen_prep(&xs, b.screen, st));
     xs.screen = b.screen;
     SKM_TRY(tc_init_stats(b.a.tc, st));
@@ -748,6 +835,9 @@ int skm_fit_hierarchical(const skm_hier_config *cfg, const skm_data *x, const in
     SKM_CUDA_TRY(cudaMemsetAsync(b.status, 0, sizeof(int), st));
     if (x->repr == SKM_REPR_RBQ1)
         SKM_CUDA_TRY(launch_rbq1_decode_rows(static_cast<const uint32_t *>(xs.x), xs.F, n, d, x->m, xs.rbq1_exp,
+                                             b.init_pos, k, static_cast<float *>(C_out), b.status, st));
+    else if (x->repr == SKM_REPR_LVQ4)
+        SKM_CUDA_TRY(launch_lvq4_decode_rows(static_cast<const uint32_t *>(xs.x), b.lvq, n, d, xs.rbq1_exp,
                                              b.init_pos, k, static_cast<float *>(C_out), b.status, st));
     else
         SKM_CUDA_TRY(launch_gather_rows(xs.x, n, x->repr == SKM_REPR_SQ8 ? 1 : 4, d, b.init_pos, k, C_out,
@@ -825,6 +915,10 @@ int skm_update_finalize(const skm_data *x, const void *partial, const int64_t *c
         SKM_CUDA_TRY(launch_finalize_rbq1(static_cast<const int64_t *>(partial), counts, k, x->d,
                                           x->m, x->rbq1_exp, static_cast<float *>(C_inout), st));
         break;
+    case SKM_REPR_LVQ4:
+        SKM_CUDA_TRY(launch_finalize_lvq4(static_cast<const int64_t *>(partial), counts, k, x->d, x->rbq1_exp,
+                                          static_cast<float *>(C_inout), st));
+        break;
     }
     return SKM_OK;
 }
@@ -866,6 +960,12 @@ int skm_fit(const skm_fit_config *cfg, const skm_data *x, const void *C_init,
         SKM_CUDA_TRY(cudaStreamSynchronize(st));
         xd.rbq1_exp = e;
     }
+    if (x->repr == SKM_REPR_LVQ4) {
+        SKM_CUDA_TRY(launch_lvq4_exponent(reinterpret_cast<const float4 *>(x->lvq), n, b.maxbits, b.e_dev, st));
+        SKM_CUDA_TRY(cudaMemcpyAsync(&e, b.e_dev, sizeof(int), cudaMemcpyDeviceToHost, st));
+        SKM_CUDA_TRY(cudaStreamSynchronize(st));
+        xd.rbq1_exp = e;
+    }
     // STEP 1: initial centroids
     SKM_CUDA_TRY(cudaMemsetAsync(b.status, 0, sizeof(int), st));
     SKM_CUDA_TRY(cudaMemsetAsync(b.u.flag, 0, sizeof(int32_t), st));
@@ -876,6 +976,10 @@ int skm_fit(const skm_fit_config *cfg, const skm_data *x, const void *C_init,
         SKM_CUDA_TRY(launch_rbq1_decode_rows(static_cast<const uint32_t *>(x->x), x->F, n, d, x->m,
                                              e, init_idx, k, static_cast<float *>(C_out), b.status,
                                              st));
+    } else if (x->repr == SKM_REPR_LVQ4) {
+        SKM_CUDA_TRY(launch_lvq4_decode_rows(static_cast<const uint32_t *>(x->x),
+                                             reinterpret_cast<const float4 *>(x->lvq), n, d, e, init_idx, k,
+                                             static_cast<float *>(C_out), b.status, st));
     } else {
         const int eb = x->repr == SKM_REPR_SQ8 ? 1 : (x->repr == SKM_REPR_BF16 ? 2 : 4);
         if (x->repr == SKM_REPR_BF16)

@@ -69,6 +69,15 @@ __device__ __forceinline__ void add_if_bit2(uint32_t &lo, uint32_t &hi, uint32_t
         : "r"(mask), "r"(flo), "r"(fhi));
 }
 
+// e4m3 encodings of the integers 0..15 (sign 0, exponent bias 7, 3 mantissa
+// bits): 0 -> 0x00, 1 -> 0x38, 2 -> 0x40, 3 -> 0x44, 4 -> 0x48, ... 15 -> 0x57.
+__device__ __forceinline__ uint8_t e4m3_of_code(uint32_t y) {
+    if (y == 0) return 0;
+    const int e = 31 - __clz(y);                // floor(log2 y), 0..3
+    const uint32_t mant = (y << (3 - e)) & 7u;  // 3 bits below the leading one
+    return (uint8_t)(((uint32_t)(e + 7) << 3) | mant);
+}
+
 // Per-centroid terms of the RBQ1 estimator (Eq. final:rabitq), one record
 // per centroid: SQ4 bias and scale multiplied by fl(1/sqrt(d)) (bd = b isd,
 // sd = s isd), the sum of codes, ||c - m||^2.
@@ -208,6 +217,41 @@ cudaError_t launch_cov_partial(const float *X, int64_t n, int d, const float *me
                                double *partial, int splits, cudaStream_t st);
 cudaError_t launch_cov_reduce(const double *partial, int splits, int d, double *cov,
                               cudaStream_t st);
+
+// LVQ4 (Section 3.1 "LVQ4"; k_lvq4.cu).  Codes: uint32 [n][ceil(d/8)] nibbles;
+// per-vector terms float4 (s, b, N, A) for points, (s, b, N, G) for centroids.
+__host__ __device__ inline int lvq4_words(int d) { return (d + 7) / 8; }
+cudaError_t launch_lvq4_encode(const float *X, int64_t n, int d, uint32_t *codes, float4 *fac,
+                               cudaStream_t st);
+cudaError_t launch_lvq4_exponent(const float4 *fac, int64_t n, unsigned int *maxbits, int *e_dev,
+                                 cudaStream_t st);
+// centroid re-encoding: yq != nullptr -> e4m3 bytes (row stride dq); yw != nullptr
+// -> nibble words; info (s, b, N, G) per centroid
+cudaError_t launch_lvq4_cprep(const float *C, int k, int d, uint8_t *yq, int dq, uint32_t *yw,
+                              float4 *info, cudaStream_t st);
+// nibble codes -> e4m3 bytes, row stride dq
+cudaError_t launch_lvq4_expand(const uint32_t *codes, int64_t n, int d, uint8_t *xs, int dq,
+                               cudaStream_t st);
+// column-pair records for the tensor epilogue: bg = (b x2, G x2), sn = (s x2, N x2)
+cudaError_t launch_lvq4_pack_pairs(const float4 *info, int k, int kp, float4 *bg, float4 *sn,
+                                   cudaStream_t st);
+cudaError_t launch_assign_lvq4_simt(const uint32_t *codes, const float4 *fac, int64_t n, int d,
+                                    const uint32_t *yw, const float4 *info, int k, int32_t *assign,
+                                    float *dist, cudaStream_t st);
+// Sq = round(s 2^e) (uint32) and Bq = round(b 2^e) (int64) in cluster-sorted order
+cudaError_t launch_lvq4_q(const float4 *fac, const int32_t *perm, const int64_t *offsets, int k, int64_t n,
+                          int e, uint32_t *sq, int64_t *bq, cudaStream_t st);
+bool ring_sum_lvq4_ok(const void *codes, int d);
+cudaError_t launch_ring_sum_lvq4(const uint32_t *codes, const uint32_t *sq, const int64_t *bq, int64_t n,
+                                 int d, const int32_t *perm, const int32_t *scl, const int64_t *offsets,
+                                 int k, int64_t *T, int32_t *flag, cudaStream_t st);
+cudaError_t launch_chunk_sum_lvq4(const uint32_t *codes, const uint32_t *sq, const int64_t *bq, int64_t n,
+                                  int d, const int32_t *perm, const int32_t *scl, const int64_t *offsets,
+                                  int k, int64_t *T, cudaStream_t st);
+cudaError_t launch_finalize_lvq4(const int64_t *partial, const int64_t *counts, int k, int d, int e,
+                                 float *C_inout, cudaStream_t st);
+cudaError_t launch_lvq4_decode_rows(const uint32_t *codes, const float4 *fac, int64_t n, int d, int e,
+                                    const int64_t *idx, int k, float *out, int *status, cudaStream_t st);
 
 // host helpers (skm_linalg.cpp)
 void philox_gaussians(uint64_t seed, int64_t count, double *out);

@@ -12,6 +12,9 @@ constexpr int TC_SQ8_MAX_D = 1024;
 // (P < 2^14) the accumulation error stays far below 1/2.  Beyond it the
 // AND + popcount kernel is used.
 constexpr int TC_RBQ1_MAX_D = 1024;
+// LVQ4 on the same e4m3 path: P <= 225 d stays below 2^18 up to this d; beyond
+// it the __dp4a kernel is used.
+constexpr int TC_LVQ4_MAX_D = 1024;
 
 struct TcAssignBufs {
     int64_t *stats = nullptr;     // [0] rescored rows, [1] fallback rows, [2] timeout (cumulative)
@@ -22,7 +25,8 @@ struct TcAssignBufs {
     float2 *cinfoz = nullptr;
     int32_t *nc = nullptr;        // SQ8: centred ||c||^2
     Rbq1CInfo *rinfo = nullptr;   // RBQ1: per-centroid estimator terms
-    float4 *rpair_bs = nullptr;   // RBQ1: the same as column-pair records (padded)
+    float4 *linfo = nullptr;      // LVQ4: per-centroid (s, b, N, G)
+    float4 *rpair_bs = nullptr;   // RBQ1 / LVQ4: column-pair records (padded)
     float4 *rpair_qn = nullptr;
     int32_t *cand = nullptr;      // F32/BF16: [n][5] screen candidates + count
     int32_t *resc_rows = nullptr;
@@ -55,6 +59,9 @@ int tc_assign_sq8(const skm_data *x, const uint8_t *C, int k, int32_t *nx_plain,
 // RBQ1 on tensor cores (e4m3 operands, exact integer P, same fp32 epilogue
 // as the AND+popcount kernel).
 int tc_assign_rbq1(const skm_data *x, const float *C, int k, int32_t *assign, float *dist,
+                   TcAssignBufs &b, cudaStream_t st, const TcSeg *seg = nullptr);
+// LVQ4 on tensor cores (e4m3 codes, exact integer P, Eq. final:lvq epilogue).
+int tc_assign_lvq4(const skm_data *x, const float *C, int k, int32_t *assign, float *dist,
                    TcAssignBufs &b, cudaStream_t st, const TcSeg *seg = nullptr);
 // Copies the cumulative statistics; returns SKM_ERR_TIMEOUT if a pipeline
 // wait gave up.  Synchronises the stream.

@@ -104,3 +104,34 @@ def test_make_rotation_is_orthogonal_and_seeded(skm):
     np.testing.assert_array_equal(P.astype(np.float32), P2)
     P3 = skm.skm_make_rotation(8, 48).numpy()
     assert not np.allclose(P2, P3)
+
+
+def test_lvq4_arguments_are_rejected_before_launch(skm):
+    L = skm.lib()
+
+    def lvq_data(n=100, d=16, lvq=0x2000):
+        x = skm.Data(skm.REPR_LVQ4, d, n, 0x1000, None, None, None, None, 0, 0)
+        x.lvq = lvq
+        return x
+
+    # the per-point terms are required and must be 16-byte aligned
+    assert L.skm_assign(ctypes.byref(lvq_data(lvq=None)), FAKE, 4, None, FAKE, None, FAKE, 1 << 30, None) == 1
+    assert L.skm_assign(ctypes.byref(lvq_data(lvq=0x2004)), FAKE, 4, None, FAKE, None, FAKE, 1 << 30, None) == 1
+    # more points than the fixed-point sums allow
+    assert L.skm_assign(ctypes.byref(lvq_data(n=(1 << 26) + 1)), FAKE, 4, None, FAKE, None, FAKE, 1 << 40,
+                        None) == 2
+    # workspace sizes exist for assign / update / fit (tensor path and the d > 1024 path)
+    for d in (16, 768, 2048):
+        for op in (0, 1, 2):
+            assert L.skm_workspace_size(op, ctypes.byref(lvq_data(d=d)), 4) > 0
+    # quantize: NULL or misaligned outputs
+    qp = skm.QuantParams(0, 0, None, None, None, None, None, None, None)
+    assert L.skm_quantize(skm.REPR_LVQ4, FAKE, 10, 16, ctypes.byref(qp), FAKE, FAKE, 1 << 20, None) == 1
+    qp.lvq = 0x2008
+    assert L.skm_quantize(skm.REPR_LVQ4, FAKE, 10, 16, ctypes.byref(qp), FAKE, FAKE, 1 << 20, None) == 1
+    # exponent: misaligned terms
+    e = ctypes.c_int(0)
+    assert L.skm_lvq4_exponent(ctypes.c_void_p(0x2004), 10, ctypes.byref(e), FAKE, 1 << 20, None) == 1
+    # hierarchical fit needs d <= 1024
+    cfg = skm.HierConfig(8, 2, 1, 1, 0)
+    assert L.skm_hier_workspace_size(ctypes.byref(cfg), ctypes.byref(lvq_data(d=2048))) == 0

@@ -721,3 +721,137 @@ def test_raw_vector_last_update_and_full_dimensional_centroids(skm):
     Cmo, _ = oracle.update_f32(X.numpy(), ap.cpu().numpy(), Cu)
     rel = np.linalg.norm(Cm.cpu().numpy() - Cmo, axis=1) / np.maximum(np.linalg.norm(Cmo, axis=1), 1e-30)
     assert rel.max() <= 1e-4
+
+
+# --------------------------------------------------------------------- LVQ4
+def _lvq4_host(q, d):
+    words = q["codes"].cpu().numpy().view(np.uint32)
+    return {"words": words, "codes": oracle.lvq4_unpack(words, d), "fac": q["lvq"].cpu().numpy()}
+
+
+@pytest.mark.parametrize("n,d", [(3000, 768), (777, 33), (500, 32), (400, 31), (100, 1), (300, 2048)])
+def test_encode_lvq4_bitexact(skm, n, d):
+    X = _points(n, d, seed=n + 3)
+    q = skm.skm_quantize(skm.REPR_LVQ4, X.to(DEV))
+    h = _lvq4_host(q, d)
+    codes, fac, _ = oracle.lvq4_encode(X.numpy())
+    np.testing.assert_array_equal(h["words"], oracle.lvq4_pack(codes))
+    np.testing.assert_array_equal(h["fac"], fac)
+
+
+@pytest.mark.parametrize("n,d,k", [(3000, 768, 300), (777, 33, 7), (500, 64, 1), (1000, 1024, 65),
+                                   (600, 1500, 40), (300, 5, 300), (2100, 128, 513)])
+def test_assign_update_lvq4_bitexact(skm, n, d, k):
+    X = _points(n, d, seed=n + 4)
+    q = skm.skm_quantize(skm.REPR_LVQ4, X.to(DEV))
+    pts = skm.lvq4_points(q, d)
+    h = _lvq4_host(q, d)
+    assert pts.rbq1_exp == oracle.lvq4_exponent(h["fac"])
+    C = X[synth.forgy_indices(n, k, seed=6)].clone()
+    a, dist = skm.skm_assign(pts, C.to(DEV))
+    ao, do = oracle.lvq4_assign(h["codes"], h["fac"], oracle.lvq4_encode(C.numpy()))
+    np.testing.assert_array_equal(a.cpu().numpy(), ao)
+    np.testing.assert_array_equal(dist.cpu().numpy(), do)
+    Cn, counts = skm.skm_update(pts, a, C.to(DEV).clone())
+    Co, co = oracle.lvq4_update(h["codes"], h["fac"], pts.rbq1_exp, ao, C.numpy())
+    np.testing.assert_array_equal(counts.cpu().numpy(), co)
+    np.testing.assert_array_equal(Cn.cpu().numpy(), Co)
+
+
+@pytest.mark.parametrize("d", [1024, 777])
+def test_assign_lvq4_large_code_products_exact(skm, d):
+    """Codes near 15 everywhere (P close to 225 d, the largest the tensor path
+    meets): the e4m3 accumulator must still give the exact integer P, seen
+    through bit-exact distances."""
+    rng = np.random.default_rng(d)
+    n, k = 700, 300
+    X = np.ones((n, d), np.float32)
+    X[np.arange(n), rng.integers(0, d, n)] = 0.0  # one code 0 per row, the rest 15
+    X[: n // 2] -= rng.integers(0, 2, (n // 2, d)).astype(np.float32) / 15.0  # codes 14 / 15 mixed
+    X[: n // 2, 0] = 0.0
+    C = np.ones((k, d), np.float32)
+    C[np.arange(k), rng.integers(0, d, k)] = 0.0
+    C[k // 2:] -= rng.integers(0, 3, (k - k // 2, d)).astype(np.float32) / 15.0
+    q = skm.skm_quantize(skm.REPR_LVQ4, torch.from_numpy(X).to(DEV))
+    pts = skm.lvq4_points(q, d)
+    h = _lvq4_host(q, d)
+    assert h["codes"].mean() > 14.0
+    a, dist = skm.skm_assign(pts, torch.from_numpy(C).to(DEV))
+    ao, do = oracle.lvq4_assign(h["codes"], h["fac"], oracle.lvq4_encode(C))
+    np.testing.assert_array_equal(a.cpu().numpy(), ao)
+    np.testing.assert_array_equal(dist.cpu().numpy(), do)
+
+
+@pytest.mark.parametrize("split", [False, True])
+def test_fit_lvq4_trajectory_bitexact(skm, split):
+    n, d, k, iters = 8000, 256, 50, 6
+    X = _points(n, d, seed=10)
+    q = skm.skm_quantize(skm.REPR_LVQ4, X.to(DEV))
+    pts = skm.lvq4_points(q, d)
+    idx = synth.forgy_indices(n, k, seed=10)
+    policy = skm.EMPTY_SPLIT if split else skm.EMPTY_KEEP
+    C, a, dist, obj, _ = skm.skm_fit(pts, k, iters, init_idx=idx.to(DEV), empty_policy=policy)
+    h = _lvq4_host(q, d)
+    C0 = oracle.lvq4_decode_points(h["codes"], h["fac"], pts.rbq1_exp, idx.numpy())
+    Co, ao = oracle.lloyd_lvq4(h["codes"], h["fac"], C0, iters, pts.rbq1_exp, split=split)
+    np.testing.assert_array_equal(a.cpu().numpy(), ao)
+    np.testing.assert_array_equal(C.cpu().numpy(), Co)
+    _, do = oracle.lvq4_assign(h["codes"], h["fac"], oracle.lvq4_encode(Co))
+    np.testing.assert_array_equal(dist.cpu().numpy(), do)
+    assert math.isclose(obj[-1], float(do.astype(np.float64).sum()), rel_tol=1e-12)
+
+
+def test_sharded_update_lvq4_matches_single(skm):
+    n, d, k = 4000, 64, 20
+    X = _points(n, d, seed=22)
+    q = skm.skm_quantize(skm.REPR_LVQ4, X.to(DEV))
+    pts = skm.lvq4_points(q, d)
+    C = X[:k].clone().to(DEV)
+    a, _ = skm.skm_assign(pts, C)
+    C_single, cnt_single = skm.skm_update(pts, a, C.clone())
+    total = torch.zeros((k, d + 1), dtype=torch.int64, device=DEV)
+    counts = torch.zeros(k, dtype=torch.int64, device=DEV)
+    for lo, hi in zip([0, 999, 1000, 3001], [999, 1000, 3001, n]):
+        part = torch.zeros((k, d + 1), dtype=torch.int64, device=DEV)
+        sp = skm.Points(skm.REPR_LVQ4, pts.x[lo:hi].contiguous(), d, rbq1_exp=pts.rbq1_exp,
+                        lvq=pts.lvq[lo:hi].contiguous())
+        skm.skm_update(sp, a[lo:hi].contiguous(), None, counts=counts, partial=part)
+        skm.skm_merge_partials(total, part)
+    C_merged = skm.skm_update_finalize(pts, total, counts, C.clone())
+    assert torch.equal(counts, cnt_single)
+    assert torch.equal(C_merged, C_single)
+
+
+def test_assign_segmented_lvq4_per_group(skm):
+    group, base = _segments()
+    n, k, d = group.size, int(base[-1]), 96
+    X = _points(n, d, seed=44)
+    Cf = _points(k, d, seed=45)
+    q = skm.skm_quantize(skm.REPR_LVQ4, X.to(DEV))
+    pts = skm.lvq4_points(q, d)
+    h = _lvq4_host(q, d)
+    a, dist = skm.skm_assign_segmented(pts, Cf.to(DEV), torch.from_numpy(group).to(DEV),
+                                       torch.from_numpy(base).to(DEV))
+    for s in range(len(_SEG_SIZES)):
+        rows = np.nonzero(group == s)[0]
+        ao, do = oracle.lvq4_assign(h["codes"][rows], h["fac"][rows],
+                                    oracle.lvq4_encode(Cf.numpy()[base[s]:base[s + 1]]))
+        np.testing.assert_array_equal(a.cpu().numpy()[rows] - base[s], ao)
+        np.testing.assert_array_equal(dist.cpu().numpy()[rows], do)
+
+
+@pytest.mark.parametrize("refine", [False, True])
+def test_fit_hierarchical_lvq4_bitexact(skm, refine):
+    n, d, k, m = 8000, 128, 48, 6
+    X = _hier_points(n, d, 53)
+    q = skm.skm_quantize(skm.REPR_LVQ4, X.to(DEV))
+    pts = skm.lvq4_points(q, d)
+    h = _lvq4_host(q, d)
+    idx = synth.forgy_indices(n, m, seed=53)
+    C, a, meso, kf, _ = skm.skm_fit_hierarchical(pts, k, m, idx.to(DEV), 3, 3, refine=refine)
+    data = {"codes": h["codes"], "fac": h["fac"], "e": pts.rbq1_exp}
+    Co, ao, amo, kfo = oracle.hierarchical("lvq4", data, k, m, idx.numpy(), 3, 3, refine=refine)
+    assert kf == kfo
+    np.testing.assert_array_equal(meso.cpu().numpy(), amo)
+    np.testing.assert_array_equal(a.cpu().numpy(), ao)
+    np.testing.assert_array_equal(C.cpu().numpy(), Co)

@@ -696,3 +696,20 @@ def test_lloyd_lvq4_points_as_centroids():
     np.testing.assert_array_equal(yc, codes)
     C, a = oracle.lloyd_lvq4(codes, fac, C0, 3, e=e)
     np.testing.assert_array_equal(a, np.arange(24))
+
+
+def test_hierarchical_lvq4_one_meso_cluster_equals_lloyd():
+    """m = 1: the fine phase is plain LVQ4 Lloyd from the evenly spaced
+    members (positions floor(t n / k))."""
+    r = _rng(47)
+    n, d, k = 600, 24, 6
+    X = r.standard_normal((n, d)).astype(np.float32)
+    codes, fac, _ = oracle.lvq4_encode(X)
+    e = oracle.lvq4_exponent(fac)
+    data = {"codes": codes, "fac": fac, "e": e}
+    C, a, am, kf = oracle.hierarchical("lvq4", data, k, 1, np.array([3]), 2, 3)
+    assert kf == [k] and np.all(am == 0)
+    init = (np.arange(k) * n) // k
+    C2, a2 = oracle.lloyd_lvq4(codes, fac, oracle.lvq4_decode_points(codes, fac, e, init), 3, e=e)
+    np.testing.assert_array_equal(C, C2)
+    np.testing.assert_array_equal(a, a2)
