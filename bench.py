@@ -485,6 +485,10 @@ def run_case(args):
         pts = skm.rbq1_points(skm.skm_quantize(skm.REPR_RBQ1, X), d)
         if args.case == "assign_rbq1":
             pts = pts.with_screen()
+    elif args.case in ("assign_lvq4", "update_lvq4"):
+        pts = skm.lvq4_points(skm.skm_quantize(skm.REPR_LVQ4, X), d)
+        if args.case == "assign_lvq4":
+            pts = pts.with_screen()
     elif args.case in ("assign_sq8", "update_sq8"):
         q = skm.skm_quantize(skm.REPR_SQ8, X)
         pts = skm.Points(skm.REPR_SQ8, q["codes"], d).with_screen()
@@ -589,6 +593,10 @@ def run_config(args):
         pR = skm.rbq1_points(q, spec.d).with_screen()
         CR, _, _, _, _ = skm.skm_fit(pR, k, 0, init_idx=idx, want_objective=False, want_dist=False)
         runs.append(("rbq1", pR, CR, spec.d, 2 * bf16_peak, "e4m3"))
+    if args.config in ("c1", "c2"):
+        pL = skm.lvq4_points(skm.skm_quantize(skm.REPR_LVQ4, X), spec.d).with_screen()
+        CL, _, _, _, _ = skm.skm_fit(pL, k, 0, init_idx=idx, want_objective=False, want_dist=False)
+        runs.append(("lvq4", pL, CL, spec.d, 2 * bf16_peak, "e4m3"))
     if args.config == "c2":
         q = skm.skm_quantize(skm.REPR_SQ8, X)
         del X
@@ -599,6 +607,10 @@ def run_config(args):
         Y = skm.skm_project(X, P)
         del X
         q = skm.skm_quantize(skm.REPR_RBQ1, Y)
+        if args.lvq4:
+            pL = skm.lvq4_points(skm.skm_quantize(skm.REPR_LVQ4, Y), spec.d).with_screen()
+            CL, _, _, _, _ = skm.skm_fit(pL, k, 0, init_idx=idx, want_objective=False, want_dist=False)
+            runs.append(("lvq4", pL, CL, spec.d, 2 * bf16_peak, "e4m3"))
         del Y
         pR = skm.rbq1_points(q, spec.d).with_screen()
         CR, _, _, _, _ = skm.skm_fit(pR, k, 0, init_idx=idx, want_objective=False, want_dist=False)
@@ -667,8 +679,8 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-popcount", action="store_true")
     ap.add_argument("--case", default=None,
-                    help="single-operation run for profiling: assign_f32|assign_rbq1|assign_sq8|"
-                         "assign_rbq1_popcount|assign_prune|update_f32|update_rbq1|update_sq8")
+                    help="single-operation run for profiling: assign_f32|assign_rbq1|assign_sq8|assign_lvq4|"
+                         "assign_rbq1_popcount|assign_prune|update_f32|update_rbq1|update_sq8|update_lvq4")
     ap.add_argument("--n", type=int, default=200_000)
     ap.add_argument("--d", type=int, default=768)
     ap.add_argument("--k", type=int, default=1000)
@@ -676,6 +688,7 @@ def main():
     ap.add_argument("--config", default=None, choices=["c0", "c1", "c2", "c3", "c4"],
                     help="per-configuration Lloyd iteration timing (median of iterations 2..iters)")
     ap.add_argument("--iters", type=int, default=10)
+    ap.add_argument("--lvq4", action="store_true", help="with --config c3: also time LVQ4 on the rotated points")
     ap.add_argument("--hier", action="store_true",
                     help="with --config: flat Lloyd fit against hierarchical k-means (m = sqrt k)")
     args = ap.parse_args()

@@ -3,19 +3,21 @@
 // decode-average of Section 3.1 "RabitQ").
 //
 // The cluster-sorted member order is cut into runs of RS_ROWS positions and
-// each of the RS_CW consumer warps of a CTA owns one run.  A producer warp
-// gathers the member rows of the CTA's runs with cp.async.bulk (global ->
-// shared, completion counted in bytes on one mbarrier per slot) into a ring
-// of slots per consumer warp, so that tens of rows per SM are in flight
-// without holding them in registers.  A consumer warp adds each row of its run
-// into register accumulators and flushes them into the cluster's global
-// accumulator with atomics whenever the cluster id changes and at the end of
-// the run; every warp has the same number of rows whatever the cluster sizes.
+// each of the RS_CW warps of a CTA owns one run.  A warp gathers the member
+// rows of its run with cp.async.bulk (global -> shared, completion counted in
+// bytes on one mbarrier per slot) into its own ring of slots, R rows per slot,
+// one copy per lane, so that a whole slot is requested by one instruction and
+// tens of rows per SM are in flight without holding them in registers.  It
+// adds each row into register accumulators, refills the slot it has just read
+// with the rows ns slots ahead, and flushes the accumulators into the
+// cluster's global accumulator with atomics whenever the cluster id changes
+// and at the end of the run; every warp has the same number of rows whatever
+// the cluster sizes.
 //
 // Every barrier wait is bounded (2 s of %globaltimer).  A wait that gives up
-// raises *flag (which skm_fit reports as SKM_ERR_TIMEOUT), the warp stops,
-// and the producer waits (bounded again) for the copies it issued before the
-// CTA returns, so no copy lands in the shared memory of a finished CTA.
+// raises *flag (which skm_fit reports as SKM_ERR_TIMEOUT), the warp stops, and
+// waits (bounded again) for the copies it issued before the CTA returns, so no
+// copy lands in the shared memory of a finished CTA.
 #include <algorithm>
 
 #include "skm_internal.cuh"
@@ -23,8 +25,8 @@
 namespace skm {
 namespace {
 
-constexpr int RS_CW = 8;                      // consumer warps per CTA
-constexpr int RS_THREADS = 32 * (RS_CW + 1);  // + one producer warp
+constexpr int RS_CW = 8;                      // warps per CTA, one run each
+constexpr int RS_THREADS = 32 * RS_CW;
 constexpr int RS_ROWS = 128;                  // sorted positions per consumer warp
 constexpr int RS_MAX_SLOTS = 16;              // ring slots per consumer warp
 constexpr int RS_RING_BYTES = 96 * 1024;      // all rings of a CTA
@@ -38,9 +40,6 @@ __device__ __forceinline__ unsigned long long gtimer() {
 }
 __device__ __forceinline__ void bar_init(uint32_t b, uint32_t count) {
     asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(b), "r"(count) : "memory");
-}
-__device__ __forceinline__ void bar_arrive(uint32_t b) {
-    asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(b) : "memory");
 }
 __device__ __forceinline__ void bar_arrive_tx(uint32_t b, uint32_t bytes) {
     asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(b), "r"(bytes)
@@ -91,110 +90,143 @@ __device__ __forceinline__ int run_len(int64_t nval, int64_t q0) {
     return r <= 0 ? 0 : (r >= RS_ROWS ? RS_ROWS : (int)r);
 }
 
-// Shared-memory layout of one CTA: ns slots per consumer warp, each holding
-// up to R rows of rb bytes (small rows are batched so that one barrier round
-// trip covers about a kilobyte).
+// Shared-memory layout of one CTA: ns slots per warp, each holding up to R
+// rows of rb bytes (R <= 32: one row per lane).
 struct RingLayout {
     int ns, R, rb;
+    int lsu;  // 1: rows gathered by 16-byte cp.async per lane (ns == LSU_STAGES)
     __host__ __device__ size_t slot_bytes() const { return (size_t)R * rb; }
     __host__ __device__ size_t ring_bytes() const { return (size_t)RS_CW * ns * slot_bytes(); }
     __host__ __device__ size_t bytes() const {
-        return ring_bytes() + (size_t)2 * RS_CW * ns * 8 + (size_t)RS_CW * RS_ROWS * 4 + 2 * RS_CW * 4;
+        return ring_bytes() + (size_t)RS_CW * ns * 8 + (size_t)RS_CW * RS_ROWS * 4;
     }
 };
 
-// Producer and teardown shared by every row type.  A consumer warp calls
-// cons.start(q0, cnt, lane) before the first row of its run (positions q0 ..
-// q0 + cnt - 1), cons.row(i, row, lane) for its i-th row (in shared memory),
-// and cons.finish(lane) after the last.
+// Gather loop shared by every row type.  A warp calls cons.start(q0, cnt,
+// lane) before the first row of its run (positions q0 .. q0 + cnt - 1),
+// cons.row(i, row, lane) for its i-th row (in shared memory), and
+// cons.finish(lane) after the last.
 template <typename Consumer>
 __device__ __forceinline__ void ring_run(const uint8_t *__restrict__ rows,
                                          const int32_t *__restrict__ perm, int64_t nval,
                                          RingLayout L, volatile int32_t *flag, Consumer &cons) {
     extern __shared__ __align__(128) uint8_t rs_smem[];
-    uint8_t *ring = rs_smem;
-    uint64_t *full = reinterpret_cast<uint64_t *>(rs_smem + L.ring_bytes());
-    uint64_t *empty = full + RS_CW * L.ns;
-    int32_t *sperm = reinterpret_cast<int32_t *>(empty + RS_CW * L.ns);
-    int32_t *issued = sperm + RS_CW * RS_ROWS;  // slots filled, per stream
-    int32_t *consumed = issued + RS_CW;         // slots released, per stream
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int64_t qbase = (int64_t)blockIdx.x * RS_CW * RS_ROWS;
-    const uint32_t rb = (uint32_t)L.rb;
     const size_t sb = L.slot_bytes();
-
-    if (threadIdx.x == 0) {
-        for (int i = 0; i < RS_CW * L.ns; ++i) {
-            bar_init(su32(full + i), 1);
-            bar_init(su32(empty + i), 1);
-        }
-        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
-    }
-    if (threadIdx.x < RS_CW) {
-        issued[threadIdx.x] = 0;
-        consumed[threadIdx.x] = 0;
-    }
-    __syncthreads();
-
-    if (warp == RS_CW) {  // ------------------------------------------ producer
-        for (int i = lane; i < RS_CW * RS_ROWS; i += 32) {
-            const int64_t q = qbase + i;
-            sperm[i] = q < nval ? perm[q] : 0;
-        }
+    uint8_t *ring = rs_smem + (size_t)warp * L.ns * sb;
+    uint64_t *full = reinterpret_cast<uint64_t *>(rs_smem + L.ring_bytes()) + warp * L.ns;
+    int32_t *sperm = reinterpret_cast<int32_t *>(rs_smem + L.ring_bytes() + (size_t)RS_CW * L.ns * 8) +
+                     warp * RS_ROWS;
+    const int64_t q0 = ((int64_t)blockIdx.x * RS_CW + warp) * RS_ROWS;
+    const int cnt = run_len(nval, q0);
+    if (cnt == 0) return;  // warp-uniform; no other warp waits on this one
+    const uint32_t rb = (uint32_t)L.rb;
+    if (lane == 0)
+        for (int s = 0; s < L.ns; ++s) bar_init(su32(full + s), 1);
+    for (int i = lane; i < cnt; i += 32) sperm[i] = perm[q0 + i];
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    __syncwarp();
+    const int nch = (cnt + L.R - 1) / L.R;  // slots' worth of rows in this run
+    // chunk j -> slot j % ns: lane 0 announces the bytes, lane r copies row r
+    auto fill = [&](int j) {
+        const int s = j % L.ns;
+        const int nr = min(L.R, cnt - j * L.R);
+        const uint32_t fb = su32(full + s);
+        if (lane == 0) bar_arrive_tx(fb, (uint32_t)nr * rb);
         __syncwarp();
-        if (lane < RS_CW) {
-            const int w = lane;
-            const int cnt = run_len(nval, qbase + (int64_t)w * RS_ROWS);
-            int j = 0, s = 0;
-            uint32_t ph = 0;
-            for (int i0 = 0; i0 < cnt; i0 += L.R, ++j) {
-                const int nr = min(L.R, cnt - i0);
-                const uint32_t fb = su32(full + w * L.ns + s);
-                if (!bar_wait(su32(empty + w * L.ns + s), ph ^ 1u, flag)) break;
-                bar_arrive_tx(fb, (uint32_t)nr * rb);
-                uint8_t *dst = ring + ((size_t)w * L.ns + s) * sb;
-                for (int r = 0; r < nr; ++r)
-                    bulk_g2s(su32(dst + (size_t)r * rb), rows + (size_t)sperm[w * RS_ROWS + i0 + r] * rb, rb, fb);
-                if (++s == L.ns) {
-                    s = 0;
-                    ph ^= 1u;
-                }
-            }
-            issued[w] = j;
+        if (lane < nr)
+            bulk_g2s(su32(ring + (size_t)s * sb + (size_t)lane * rb),
+                     rows + (size_t)sperm[j * L.R + lane] * rb, rb, fb);
+    };
+    const int pre = nch < L.ns ? nch : L.ns;
+    for (int j = 0; j < pre; ++j) fill(j);
+    int issued = pre, j = 0;
+    cons.start(q0, cnt, lane);
+    for (; j < nch; ++j) {
+        const int s = j % L.ns;
+        const bool ok = bar_wait(su32(full + s), (uint32_t)(j / L.ns) & 1u, flag);
+        if (!__all_sync(0xffffffffu, ok)) break;
+        const uint8_t *src = ring + (size_t)s * sb;
+        const int nr = min(L.R, cnt - j * L.R);
+        for (int r = 0; r < nr; ++r) cons.row(j * L.R + r, src + (size_t)r * rb, lane);
+        if (j + L.ns < nch) {
+            // the slot's generic-proxy reads are ordered before the async copies
+            // that overwrite it
+            asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+            __syncwarp();
+            fill(j + L.ns);
+            ++issued;
         }
-    } else {  // ------------------------------------------------------ consumers
-        const int w = warp;
-        const int cnt = run_len(nval, qbase + (int64_t)w * RS_ROWS);
-        int j = 0;
-        if (cnt > 0) {
-            cons.start(qbase + (int64_t)w * RS_ROWS, cnt, lane);
-            int s = 0;
-            uint32_t ph = 0;
-            for (int i0 = 0; i0 < cnt; i0 += L.R, ++j) {
-                const int nr = min(L.R, cnt - i0);
-                const bool ok = bar_wait(su32(full + w * L.ns + s), ph, flag);
-                if (!__all_sync(0xffffffffu, ok)) break;
-                const uint8_t *src = ring + ((size_t)w * L.ns + s) * sb;
-                for (int r = 0; r < nr; ++r) cons.row(i0 + r, src + (size_t)r * rb, lane);
-                __syncwarp();
-                if (lane == 0) bar_arrive(su32(empty + w * L.ns + s));
-                if (++s == L.ns) {
-                    s = 0;
-                    ph ^= 1u;
-                }
-            }
-            cons.finish(lane);
-        }
-        if (lane == 0) consumed[w] = j;
     }
-    __syncthreads();
-    // slots filled but never released (only after a wait gave up): let their
+    cons.finish(lane);
+    // slots filled but never read (only after a wait gave up): let their
     // copies land before the CTA's shared memory goes away
-    if (warp == RS_CW && lane < RS_CW) {
-        const int w = lane;
-        for (int j = consumed[w]; j < issued[w]; ++j)
-            if (!bar_wait_drain(su32(full + w * L.ns + j % L.ns), (uint32_t)(j / L.ns) & 1u)) break;
+    for (int jj = j; jj < issued; ++jj)
+        if (!bar_wait_drain(su32(full + jj % L.ns), (uint32_t)(jj / L.ns) & 1u)) break;
+    __syncwarp();
+}
+
+// Mid-size rows (about 1 KB, where the consumer does little work per byte):
+// the warp's lanes gather the rows themselves with 16-byte cp.async (LSU
+// path) into LSU_STAGES slots of R rows, one commit group per slot; a
+// slot is read once cp.async.wait_group leaves only the younger groups
+// pending (empty groups keep the count uniform at the tail).  These loads
+// always complete, so there is no wait that could hang.
+constexpr int LSU_STAGES = 4;
+template <typename Consumer>
+__device__ __forceinline__ void ring_run_lsu(const uint8_t *__restrict__ rows,
+                                             const int32_t *__restrict__ perm, int64_t nval,
+                                             RingLayout L, Consumer &cons) {
+    extern __shared__ __align__(128) uint8_t rs_smem[];
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const size_t sb = L.slot_bytes();
+    uint8_t *ring = rs_smem + (size_t)warp * LSU_STAGES * sb;
+    int32_t *sperm = reinterpret_cast<int32_t *>(rs_smem + L.ring_bytes() + (size_t)RS_CW * L.ns * 8) +
+                     warp * RS_ROWS;
+    const int64_t q0 = ((int64_t)blockIdx.x * RS_CW + warp) * RS_ROWS;
+    const int cnt = run_len(nval, q0);
+    if (cnt == 0) return;
+    for (int i = lane; i < cnt; i += 32) sperm[i] = perm[q0 + i];
+    __syncwarp();
+    const int rb = L.rb, per_row = rb >> 4;  // 16-byte pieces per row
+    const int nch = (cnt + L.R - 1) / L.R;
+    auto fill = [&](int j) {  // always commits one group (empty past the last chunk)
+        if (j < nch) {
+            uint8_t *dst = ring + (size_t)(j % LSU_STAGES) * sb;
+            const int nr = min(L.R, cnt - j * L.R);
+            for (int r = 0; r < nr; ++r) {
+                const uint8_t *src = rows + (size_t)sperm[j * L.R + r] * rb;
+                for (int c = lane; c < per_row; c += 32)
+                    asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(su32(dst + (size_t)r * rb + 16 * c)),
+                                 "l"(src + 16 * c)
+                                 : "memory");
+            }
+        }
+        asm volatile("cp.async.commit_group;" ::: "memory");
+    };
+#pragma unroll
+    for (int j = 0; j < LSU_STAGES; ++j) fill(j);
+    cons.start(q0, cnt, lane);
+    for (int j = 0; j < nch; ++j) {
+        asm volatile("cp.async.wait_group %0;" ::"n"(LSU_STAGES - 1) : "memory");
+        __syncwarp();
+        const uint8_t *src = ring + (size_t)(j % LSU_STAGES) * sb;
+        const int nr = min(L.R, cnt - j * L.R);
+        for (int r = 0; r < nr; ++r) cons.row(j * L.R + r, src + (size_t)r * rb, lane);
+        __syncwarp();  // every lane has read the slot before it is refilled
+        fill(j + LSU_STAGES);
     }
+    cons.finish(lane);
+    asm volatile("cp.async.wait_group 0;" ::: "memory");
+}
+
+template <typename Consumer>
+__device__ __forceinline__ void ring_gather(const uint8_t *__restrict__ rows, const int32_t *__restrict__ perm,
+                                            int64_t nval, RingLayout L, volatile int32_t *flag, Consumer &cons) {
+    if (L.lsu)
+        ring_run_lsu(rows, perm, nval, L, cons);
+    else
+        ring_run(rows, perm, nval, L, flag, cons);
 }
 
 // ---------------------------------------------------------- fp32 / bf16 rows
@@ -276,7 +308,7 @@ __global__ void __launch_bounds__(RS_THREADS) ring_sum_float_kernel(
     cons.S = S;
     cons.stride = stride;
     cons.d = d;
-    ring_run(static_cast<const uint8_t *>(X), perm, nval, L, flag, cons);
+    ring_gather(static_cast<const uint8_t *>(X), perm, nval, L, flag, cons);
 }
 
 // ------------------------------------------------------------- 1-bit rows
@@ -368,7 +400,7 @@ __global__ void __launch_bounds__(RS_THREADS) ring_sum_rbq1_kernel(
     cons.fqs = fqs;
     cons.T = T;
     cons.d = d;
-    ring_run(reinterpret_cast<const uint8_t *>(codes), perm, nval, L, flag, cons);
+    ring_gather(reinterpret_cast<const uint8_t *>(codes), perm, nval, L, flag, cons);
 }
 
 // --------------------------------------------------------------- SQ8 rows
@@ -455,7 +487,7 @@ __global__ void __launch_bounds__(RS_THREADS) ring_sum_sq8_kernel(
     cons.scl = scl;
     cons.S = S;
     cons.d = d;
-    ring_run(codes, perm, nval, L, flag, cons);
+    ring_gather(codes, perm, nval, L, flag, cons);
 }
 
 // ------------------------------------------------------------- LVQ4 rows
@@ -550,13 +582,27 @@ __global__ void __launch_bounds__(RS_THREADS) ring_sum_lvq4_kernel(
     cons.T = T;
     cons.d = d;
     cons.W = lvq4_words(d);
-    ring_run(reinterpret_cast<const uint8_t *>(codes), perm, nval, L, flag, cons);
+    ring_gather(reinterpret_cast<const uint8_t *>(codes), perm, nval, L, flag, cons);
 }
+
+// Rows of [RS_LSU_MIN_ROW, RS_LSU_MAX_ROW) bytes take the LSU path (per-lane
+// cp.async), all others one bulk copy each (measured on GB300 at 1M points:
+// 1 KB SQ8 rows 0.294 vs 0.331 ms per update with the LSU path; 96-512 B code
+// rows and 3 KB fp32 rows equal or faster with bulk copies).
+constexpr uint32_t RS_LSU_MIN_ROW = 1024;
+constexpr uint32_t RS_LSU_MAX_ROW = 2048;
 
 bool ring_layout(uint32_t rb, RingLayout &L) {
     if (rb == 0 || rb % 16 != 0) return false;
     L.rb = (int)rb;
-    L.R = (int)std::max<uint32_t>(1u, std::min<uint32_t>(8u, 1024u / rb));
+    if (rb >= RS_LSU_MIN_ROW && rb < RS_LSU_MAX_ROW) {
+        L.lsu = 1;
+        L.ns = LSU_STAGES;
+        L.R = (int)std::max<size_t>(1, std::min<size_t>(32, RS_RING_BYTES / ((size_t)RS_CW * LSU_STAGES * rb)));
+        return true;
+    }
+    L.lsu = 0;
+    L.R = (int)std::max<uint32_t>(1u, std::min<uint32_t>(32u, 2048u / rb));
     L.ns = (int)std::min<size_t>(RS_MAX_SLOTS, RS_RING_BYTES / ((size_t)RS_CW * L.slot_bytes()));
     return L.ns >= 2;
 }
