@@ -493,6 +493,10 @@ def run_case(args):
         q = skm.skm_quantize(skm.REPR_SQ8, X)
         pts = skm.Points(skm.REPR_SQ8, q["codes"], d).with_screen()
         C = q["codes"][:k].clone()
+    elif args.case == "assign_prune_sq8":  # SQ8 codes, exact integer prefix-block pruning
+        q = skm.skm_quantize(skm.REPR_SQ8, X)
+        pts = skm.Points(skm.REPR_SQ8, q["codes"], d, flags=skm.FLAG_PRUNE)
+        C = q["codes"][synth.forgy_indices(n, k, seed=0).cuda()].clone()
     elif args.case == "assign_prune":  # bf16 points, exact prefix-block pruning
         Xb = X.to(torch.bfloat16).view(torch.int16).contiguous()
         pts = skm.Points(skm.REPR_BF16, Xb, d, flags=skm.FLAG_PRUNE)
@@ -602,6 +606,9 @@ def run_config(args):
         del X
         runs.append(("sq8", skm.Points(skm.REPR_SQ8, q["codes"], spec.d).with_screen(),
                      q["codes"][idx].clone(), spec.d, bf16_peak, "bf16"))
+        if args.prune:
+            runs.append(("sq8_prune", skm.Points(skm.REPR_SQ8, q["codes"], spec.d, flags=skm.FLAG_PRUNE),
+                         q["codes"][idx].clone(), spec.d, None, "int32 CUDA cores"))
     if args.config == "c3":
         P = synth.haar_rotation(spec.d, 99).to(torch.float32).contiguous().to(dev)
         Y = skm.skm_project(X, P)
@@ -647,7 +654,7 @@ def run_config(args):
             torch.cuda.synchronize()
             ta.append(e0.elapsed_time(e1))
             tu.append(e1.elapsed_time(e2))
-            if label == "bf16_prune":
+            if label.endswith("_prune"):
                 prev = a.clone()
         sel = slice(1, None) if iters > 1 else slice(0, None)
         t_a = float(np.median(ta[sel]))
@@ -660,7 +667,7 @@ def run_config(args):
             ach = 2.0 * n * k * d / (t_a / 1e3) / 1e12
             out["assign_roofline"] = {"bound": "tensor", "achieved_tflops": round(ach, 2),
                                       "peak_tflops": peak, "frac": round(ach / peak, 4), "flop": kind}
-        if label == "bf16_prune":
+        if label.endswith("_prune"):
             _, _, _, _, st = skm.skm_fit(pts, k, 1, C_init=C, want_objective=False, want_dist=False)
             out["prune_stats_2_assigns"] = st
             out["dense_equiv_tensor_ms"] = round(2.0 * n * k * d / (bf16_peak * 1e12) * 1e3, 3)
@@ -680,7 +687,8 @@ def main():
     ap.add_argument("--no-popcount", action="store_true")
     ap.add_argument("--case", default=None,
                     help="single-operation run for profiling: assign_f32|assign_rbq1|assign_sq8|assign_lvq4|"
-                         "assign_rbq1_popcount|assign_prune|update_f32|update_rbq1|update_sq8|update_lvq4")
+                         "assign_rbq1_popcount|assign_prune|assign_prune_sq8|update_f32|update_rbq1|update_sq8|"
+                         "update_lvq4")
     ap.add_argument("--n", type=int, default=200_000)
     ap.add_argument("--d", type=int, default=768)
     ap.add_argument("--k", type=int, default=1000)
@@ -689,6 +697,7 @@ def main():
                     help="per-configuration Lloyd iteration timing (median of iterations 2..iters)")
     ap.add_argument("--iters", type=int, default=10)
     ap.add_argument("--lvq4", action="store_true", help="with --config c3: also time LVQ4 on the rotated points")
+    ap.add_argument("--prune", action="store_true", help="with --config c2: also time SQ8 with exact pruning")
     ap.add_argument("--hier", action="store_true",
                     help="with --config: flat Lloyd fit against hierarchical k-means (m = sqrt k)")
     args = ap.parse_args()

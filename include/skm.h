@@ -65,11 +65,13 @@ typedef enum skm_dtype { SKM_DTYPE_F32 = 0, SKM_DTYPE_BF16 = 1 } skm_dtype;
 
 /* skm_data.flags */
 enum {
-    /* F32 / BF16, d <= 1024: assign by exact dimension pruning on CUDA cores
-     * (Section 3.1 "SuperKMeans": partial distances over 32-dimension prefix
-     * blocks, a centroid is dropped as soon as its partial distance exceeds
-     * the row's current best) instead of the tensor-core screen.  Same
-     * result (the fp32 nearest centroid). */
+    /* F32 / BF16 / SQ8, d <= 1024: assign by exact dimension pruning on CUDA
+     * cores (Section 3.1 "SuperKMeans", extended to SQ8 codes as the section
+     * describes: partial distances over 32-dimension prefix blocks, a
+     * centroid is dropped as soon as its partial distance exceeds the row's
+     * current best) instead of the tensor-core path.  Same result (the fp32
+     * nearest centroid; for SQ8 the exact integer code-space nearest, with
+     * integer partial sums). */
     SKM_FLAG_PRUNE = 1
 };
 

@@ -1,6 +1,7 @@
 // Exact dimension pruning (Section 3.1 "SuperKMeans": partial distances over
 // prefix blocks of the projected dimensions; a centroid is dropped once its
-// partial distance exceeds the row's current best).  CUDA cores, fp32.
+// partial distance exceeds the row's current best).  CUDA cores, fp32 (points
+// fp32 or bf16, centroids fp32) or exact integers (SQ8 codes).
 //
 // One warp per point row.  The bound beta starts at the exact distance to a
 // seed centroid (the previous assignment when given, else centroid 0).
@@ -162,7 +163,139 @@ __global__ void __launch_bounds__(PR_WARPS * 32) prune_assign_kernel(
     }
 }
 
+// ---------------------------------------------------------------- SQ8 codes
+// The same pruning on SQ8 codes (Section 3.1: SuperKMeans extended to SQ8):
+// partial distances are exact integers, sum over a 32-dimension block of
+// (xbar_i - cbar_i)^2 as |x - c| per byte (__vabsdiffu4) squared and summed by
+// __dp4a, so a centroid is dropped exactly when its partial exceeds beta (no
+// slack) and the result is the exact code-space argmin.  Point codes are
+// staged as 32-bit words (d % 4 == 0) or bytes.
+__device__ __forceinline__ int32_t block_partial_u8(const uint8_t *sx, const uint8_t *c, int d, int b, bool words) {
+    const int i0 = 32 * b;
+    int32_t s = 0;
+    if (words && i0 + 32 <= d) {
+        const uint32_t *xw = reinterpret_cast<const uint32_t *>(sx + i0);
+        const uint32_t *cw = reinterpret_cast<const uint32_t *>(c + i0);
+#pragma unroll
+        for (int q = 0; q < 8; ++q) {
+            const uint32_t df = __vabsdiffu4(xw[q], __ldg(cw + q));
+            s = (int32_t)__dp4a(df, df, (uint32_t)s);
+        }
+    } else {
+        const int i1 = min(d, i0 + 32);
+        for (int i = i0; i < i1; ++i) {
+            const int32_t t = (int32_t)sx[i] - (int32_t)__ldg(c + i);
+            s += t * t;
+        }
+    }
+    return s;
+}
+
+__global__ void __launch_bounds__(PR_WARPS * 32) prune_assign_sq8_kernel(
+    const uint8_t *__restrict__ X, int64_t n, int d, const uint8_t *__restrict__ C, int k,
+    const int32_t *__restrict__ prev, int32_t *__restrict__ assign, float *__restrict__ dist,
+    unsigned long long *__restrict__ counters) {
+    __shared__ __align__(16) uint8_t sx_all[PR_WARPS][PR_MAX_D];
+    __shared__ int qid[PR_WARPS][2][PR_BATCH];
+    __shared__ int32_t qps[PR_WARPS][2][PR_BATCH];
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const unsigned lt = (1u << lane) - 1u;
+    uint8_t *sx = sx_all[warp];
+    const int nb = (d + 31) >> 5;
+    const bool words = (d % 4) == 0 && (reinterpret_cast<uintptr_t>(C) & 3) == 0;
+    const int64_t nw = (int64_t)gridDim.x * PR_WARPS;
+    unsigned long long first_alive = 0, complete = 0;
+    for (int64_t row = (int64_t)blockIdx.x * PR_WARPS + warp; row < n; row += nw) {
+        __syncwarp();
+        for (int i = lane; i < d; i += 32) sx[i] = __ldg(X + row * d + i);
+        __syncwarp();
+        int best = prev ? prev[row] : 0;
+        if (best < 0 || best >= k) best = 0;
+        int32_t beta = 0;
+        for (int b = 0; b < nb; ++b) beta += block_partial_u8(sx, C + (int64_t)best * d, d, b, words);
+        for (int c0 = 0; c0 < k; c0 += PR_BATCH) {
+            __syncwarp();
+            int cnt = 0;
+            for (int s = 0; s < PR_BATCH / 32; ++s) {
+                const int j = c0 + 32 * s + lane;
+                const int32_t p = (j < k) ? block_partial_u8(sx, C + (int64_t)j * d, d, 0, words) : INT32_MAX;
+                const bool alive = j < k && p <= beta;
+                const unsigned m = __ballot_sync(0xffffffffu, alive);
+                if (alive) {
+                    const int pos = cnt + __popc(m & lt);
+                    qid[warp][0][pos] = j;
+                    qps[warp][0][pos] = p;
+                }
+                cnt += __popc(m);
+            }
+            first_alive += cnt;
+            int src = 0;
+            for (int b = 1; b < nb && cnt > 0; ++b) {
+                __syncwarp();
+                int ncnt = 0;
+                for (int t0 = 0; t0 < cnt; t0 += 32) {
+                    const int t = t0 + lane;
+                    const bool valid = t < cnt;
+                    const int j = valid ? qid[warp][src][t] : 0;
+                    const int32_t p = valid ? qps[warp][src][t] + block_partial_u8(sx, C + (int64_t)j * d, d, b, words) : 0;
+                    const bool alive = valid && p <= beta;
+                    const unsigned m = __ballot_sync(0xffffffffu, alive);
+                    if (alive) {
+                        const int pos = ncnt + __popc(m & lt);
+                        qid[warp][src ^ 1][pos] = j;
+                        qps[warp][src ^ 1][pos] = p;
+                    }
+                    ncnt += __popc(m);
+                }
+                cnt = ncnt;
+                src ^= 1;
+            }
+            __syncwarp();
+            complete += cnt;
+            for (int t0 = 0; t0 < cnt; t0 += 32) {
+                const int t = t0 + lane;
+                int32_t p = INT32_MAX;
+                int j = 0x7fffffff;
+                if (t < cnt) {
+                    p = qps[warp][src][t];
+                    j = qid[warp][src][t];
+                }
+#pragma unroll
+                for (int o = 16; o > 0; o >>= 1) {
+                    const int32_t op = __shfl_xor_sync(0xffffffffu, p, o);
+                    const int oj = __shfl_xor_sync(0xffffffffu, j, o);
+                    if (op < p || (op == p && oj < j)) {
+                        p = op;
+                        j = oj;
+                    }
+                }
+                if (p < beta || (p == beta && j < best)) {
+                    beta = p;
+                    best = j;
+                }
+            }
+        }
+        if (lane == 0) {
+            assign[row] = best;
+            if (dist) dist[row] = (float)beta;
+        }
+    }
+    if (counters && lane == 0) {
+        atomicAdd(&counters[0], first_alive);
+        atomicAdd(&counters[1], complete);
+    }
+}
+
 }  // namespace
+
+cudaError_t launch_prune_assign_sq8(const uint8_t *X, int64_t n, int d, const uint8_t *C, int k, const int32_t *prev,
+                                    int32_t *assign, float *dist, unsigned long long *counters, cudaStream_t st) {
+    if (n == 0) return cudaSuccess;
+    int64_t blocks = (n + PR_WARPS - 1) / PR_WARPS;
+    if (blocks > 152 * 16) blocks = 152 * 16;
+    prune_assign_sq8_kernel<<<(int)blocks, PR_WARPS * 32, 0, st>>>(X, n, d, C, k, prev, assign, dist, counters);
+    return launched();
+}
 
 cudaError_t launch_prune_assign(const void *X, int x_is_bf16, int64_t n, int d, const float *C,
                                 int k, const int32_t *prev, int32_t *assign, float *dist,

@@ -51,8 +51,8 @@ static int check_data(const skm_data *x, bool need_codes = true) {
         return set_error(x->n < 1 ? SKM_ERR_INVALID_ARG : SKM_ERR_UNSUPPORTED,
                          "n = %lld outside [1, 2^31)", (long long)x->n);
     if (need_codes && !x->x) return set_error(SKM_ERR_INVALID_ARG, "x->x is NULL");
-    if ((x->flags & SKM_FLAG_PRUNE) && (x->repr == SKM_REPR_F32 || x->repr == SKM_REPR_BF16) &&
-        x->d > PRUNE_MAX_D)
+    if ((x->flags & SKM_FLAG_PRUNE) &&
+        (x->repr == SKM_REPR_F32 || x->repr == SKM_REPR_BF16 || x->repr == SKM_REPR_SQ8) && x->d > PRUNE_MAX_D)
         return set_error(SKM_ERR_UNSUPPORTED, "SKM_FLAG_PRUNE supports d <= %d", PRUNE_MAX_D);
     if (x->repr == SKM_REPR_RBQ1) {
         if (x->n > MAX_N_RBQ1)
@@ -82,7 +82,8 @@ static int check_k(const skm_data *x, int k, bool k_le_n = false) {
 
 // ------------------------------------------------------------ workspace plans
 static bool use_prune(const skm_data *x) {
-    return (x->flags & SKM_FLAG_PRUNE) && (x->repr == SKM_REPR_F32 || x->repr == SKM_REPR_BF16);
+    return (x->flags & SKM_FLAG_PRUNE) &&
+           (x->repr == SKM_REPR_F32 || x->repr == SKM_REPR_BF16 || x->repr == SKM_REPR_SQ8);
 }
 
 struct AssignBufs {
@@ -209,9 +210,13 @@ static int do_assign(const skm_data *x, const void *C, int k, const int32_t *pre
     const int64_t n = x->n;
     const int d = x->d;
     if (use_prune(x)) {
-        SKM_CUDA_TRY(launch_prune_assign(x->x, x->repr == SKM_REPR_BF16, n, d,
-                                         static_cast<const float *>(C), k, prev, assign, dist,
-                                         b.prune, st));
+        if (x->repr == SKM_REPR_SQ8)
+            SKM_CUDA_TRY(launch_prune_assign_sq8(static_cast<const uint8_t *>(x->x), n, d, static_cast<const uint8_t *>(C),
+                                                 k, prev, assign, dist, b.prune, st));
+        else
+            SKM_CUDA_TRY(launch_prune_assign(x->x, x->repr == SKM_REPR_BF16, n, d,
+                                             static_cast<const float *>(C), k, prev, assign, dist,
+                                             b.prune, st));
         return SKM_OK;
     }
     switch (x->repr) {

@@ -129,6 +129,8 @@ cudaError_t launch_assign_exact_rows(const void *X, int x_is_bf16, const int32_t
 cudaError_t launch_prune_assign(const void *X, int x_is_bf16, int64_t n, int d, const float *C,
                                 int k, const int32_t *prev, int32_t *assign, float *dist,
                                 unsigned long long *counters, cudaStream_t st);
+cudaError_t launch_prune_assign_sq8(const uint8_t *X, int64_t n, int d, const uint8_t *C, int k, const int32_t *prev,
+                                    int32_t *assign, float *dist, unsigned long long *counters, cudaStream_t st);
 cudaError_t launch_assign_sq8_simt(const uint8_t *X, int64_t n, int d, const uint8_t *C, int k,
                                    const int32_t *nx, const int32_t *nc, int32_t *assign,
                                    float *dist, cudaStream_t st);

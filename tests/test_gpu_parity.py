@@ -855,3 +855,37 @@ def test_fit_hierarchical_lvq4_bitexact(skm, refine):
     np.testing.assert_array_equal(meso.cpu().numpy(), amo)
     np.testing.assert_array_equal(a.cpu().numpy(), ao)
     np.testing.assert_array_equal(C.cpu().numpy(), Co)
+
+
+# ------------------------------------------------- SQ8 with exact pruning
+@pytest.mark.parametrize("n,d,k", [(3000, 256, 300), (777, 33, 13), (500, 1024, 40), (2000, 64, 1)])
+def test_prune_sq8_bitexact_and_seed_independent(skm, n, d, k):
+    """SuperKMeans on SQ8 codes: integer partial distances make the pruning
+    exact, so the result is the oracle's code-space argmin bit for bit,
+    whatever seeds the bound."""
+    X = _points(n, d, seed=n + d)
+    q = skm.skm_quantize(skm.REPR_SQ8, X.to(DEV))
+    codes = q["codes"].cpu().numpy()
+    Cc = q["codes"][synth.forgy_indices(n, k, seed=8).to(DEV)].clone()
+    ao, bo = oracle.assign_sq8(codes, Cc.cpu().numpy())
+    pp = skm.Points(skm.REPR_SQ8, q["codes"], d, flags=skm.FLAG_PRUNE)
+    a0, d0 = skm.skm_assign(pp, Cc)
+    np.testing.assert_array_equal(a0.cpu().numpy(), ao)
+    np.testing.assert_array_equal(d0.cpu().numpy(), bo.astype(np.float32))
+    prev = torch.randint(0, k, (n,), generator=torch.Generator().manual_seed(9), dtype=torch.int32).to(DEV)
+    a1, d1 = skm.skm_assign(pp, Cc, prev_assign=prev)
+    assert torch.equal(a1, a0) and torch.equal(d1, d0)
+
+
+def test_prune_fit_sq8_trajectory_bitexact(skm):
+    n, d, k, iters = 6000, 128, 40, 5
+    X = _points(n, d, seed=34)
+    q = skm.skm_quantize(skm.REPR_SQ8, X.to(DEV))
+    codes = q["codes"].cpu().numpy()
+    idx = synth.forgy_indices(n, k, seed=34)
+    pp = skm.Points(skm.REPR_SQ8, q["codes"], d, flags=skm.FLAG_PRUNE)
+    C, a, _, _, st = skm.skm_fit(pp, k, iters, init_idx=idx.to(DEV))
+    Co, ao = oracle.lloyd_sq8(codes, codes[idx.numpy()], iters)
+    np.testing.assert_array_equal(a.cpu().numpy(), ao)
+    np.testing.assert_array_equal(C.cpu().numpy(), Co)
+    assert 0 < st["prune_complete"] <= st["prune_first_block"] <= (iters + 1) * n * k
