@@ -27,12 +27,14 @@
 //    an integer below 2^24 for d <= 1024, so the fp32 accumulator holds the
 //    exact integer dot product; the epilogue forms the integer distance and
 //    keeps the argmin (ties to the lowest index).
-//  RBQ1: point bits as e4m3 {0, 1} and centroid SQ4 codes as e4m3 {0..15}
-//    (kind::f8f6f4, K = 32 per instruction); the nearest integer to the
-//    accumulator is P = sum_i xbar_i ybar_i of Eq. final:rabitq (d <= 1024
-//    keeps P < 2^14 and the accumulation error far below 1/2), and the
-//    epilogue evaluates the estimator in fp32 in the library's fixed order,
-//    so the result equals the AND+popcount kernel's bit for bit.
+//  RBQ1: point bits as e4m3 -1 / +1 (2 xbar - 1) and centroid SQ4 codes as
+//    e4m3 {0..15} (kind::f8f6f4, K = 32 per instruction), so the accumulator
+//    is the exact integer 2P - sum ybar of Eq. final:rabitq (|.| <= 15 d; the
+//    products are exact and every partial sum is an integer far below 2^24),
+//    and the epilogue evaluates the estimator in fp32 in the library's fixed
+//    order, so the result equals the AND+popcount kernel's bit for bit.
+//  LVQ4: point and centroid codes 0..15 in e4m3, the accumulator is the exact
+//    integer P = <xbar, ybar> (<= 225 d) of Eq. final:lvq.
 #include <cuda.h>
 #include <cudaTypedefs.h>
 
@@ -257,6 +259,26 @@ __device__ __forceinline__ void tmem_ld32(uint32_t taddr, uint32_t (&v)[32]) {
         : "r"(taddr)
         : "memory");
     asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+}
+
+// 16 columns, no wait: the registers are valid only after tmem_wait16 on the
+// same array (which names them as operands, so nothing reads them earlier).
+__device__ __forceinline__ void tmem_ld16_async(uint32_t taddr, uint32_t (&v)[16]) {
+    asm volatile(
+        "tcgen05.ld.sync.aligned.32x32b.x16.b32 "
+        "{%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15}, [%16];"
+        : "=r"(v[0]), "=r"(v[1]), "=r"(v[2]), "=r"(v[3]), "=r"(v[4]), "=r"(v[5]), "=r"(v[6]), "=r"(v[7]),
+          "=r"(v[8]), "=r"(v[9]), "=r"(v[10]), "=r"(v[11]), "=r"(v[12]), "=r"(v[13]), "=r"(v[14]), "=r"(v[15])
+        : "r"(taddr)
+        : "memory");
+}
+__device__ __forceinline__ void tmem_wait16(uint32_t (&v)[16]) {
+    asm volatile("tcgen05.wait::ld.sync.aligned;"
+                 : "+r"(v[0]), "+r"(v[1]), "+r"(v[2]), "+r"(v[3]), "+r"(v[4]), "+r"(v[5]), "+r"(v[6]), "+r"(v[7]),
+                   "+r"(v[8]), "+r"(v[9]), "+r"(v[10]), "+r"(v[11]), "+r"(v[12]), "+r"(v[13]), "+r"(v[14]),
+                   "+r"(v[15])
+                 :
+                 : "memory");
 }
 
 // Packed fp32 pairs (two IEEE round-to-nearest operations per instruction).
@@ -612,6 +634,83 @@ __global__ void __launch_bounds__(tc_threads<NH>(), 1)
                 const uint8_t *rbuf = rec_base + b * REC_BYTES;
                 const uint32_t taddr = tmem + ((uint32_t)(q * 32) << 16) + b * BN + slice * SW;
                 const int jh = ct * BN + slice * SW;
+                if (f8_mode<MODE>()) {
+                    // e4m3 modes: 16-column chunks, the next chunk's TMEM load in
+                    // flight while this one is evaluated (two 16-register buffers)
+                    constexpr int NC = SW / 16;
+                    uint32_t va[16], vb[16];
+                    auto chunk = [&](const uint32_t(&v)[16], int c) {
+                        const int j0 = jh + c * 16;
+                        const int cc = slice * SW + c * 16;
+                        float gb[2];
+                        int gi[2];
+#pragma unroll
+                        for (int g = 0; g < 2; ++g) {
+                            gb[g] = INFINITY;
+                            gi[g] = 0x7fffffff;
+#pragma unroll
+                            for (int i = 8 * g; i < 8 * g + 8; i += 2) {
+                                const float4 r0 = reinterpret_cast<const float4 *>(rbuf)[(cc + i) >> 1];
+                                const float4 r1 = reinterpret_cast<const float4 *>(rbuf)[128 + ((cc + i) >> 1)];
+                                // the accumulator is the exact integer dot product (LVQ4:
+                                // P = <xbar, ybar>; 1-bit: 2P - sum ybar, from +-1 codes)
+                                const float2 P2 = make_float2(__uint_as_float(v[i]), __uint_as_float(v[i + 1]));
+                                float2 est;
+                                if (MODE == MODE_LVQ4) {
+                                    // Eq. final:lvq: key = fma(b_y, -2 A_x, N_y),
+                                    // fma(G_y, -2 b_x, .), fma(-2 s_x, s_y P, .)
+                                    est = ffma2(make_float2(r0.x, r0.y), make_float2(a2, a2), make_float2(r1.z, r1.w));
+                                    est = ffma2(make_float2(r0.z, r0.w), make_float2(rf2, rf2), est);
+                                    const float2 t = fmul2(make_float2(r1.x, r1.y), P2);
+                                    est = ffma2(make_float2(rpc, rpc), t, est);
+                                } else {
+                                    // Eq. final:rabitq in Eq. rabitq_l2: u = fma(sd, 2P -
+                                    // sum ybar, bd pc), est = fma(-2F, u, nx2 + ny2)
+                                    const float2 t = fmul2(make_float2(r0.x, r0.y), make_float2(rpc, rpc));
+                                    const float2 u = ffma2(make_float2(r0.z, r0.w), P2, t);
+                                    const float2 nn = fadd2(make_float2(rnx2, rnx2), make_float2(r1.z, r1.w));
+                                    est = ffma2(make_float2(rf2, rf2), u, nn);
+                                }
+                                if (SEG && (j0 < cb || j0 + 16 > ce)) {  // columns outside the row's group
+                                    if (j0 + i < cb || j0 + i >= ce) est.x = INFINITY;
+                                    if (j0 + i + 1 < cb || j0 + i + 1 >= ce) est.y = INFINITY;
+                                }
+                                if (est.x < gb[g]) {
+                                    gb[g] = est.x;
+                                    gi[g] = j0 + i;
+                                }
+                                if (est.y < gb[g]) {
+                                    gb[g] = est.y;
+                                    gi[g] = j0 + i + 1;
+                                }
+                            }
+                        }
+                        // the two groups hold increasing columns: the earlier wins ties
+#pragma unroll
+                        for (int g = 0; g < 2; ++g)
+                            if (gb[g] < fbest) {
+                                fbest = gb[g];
+                                besti = gi[g];
+                            }
+                    };
+                    if (jh < p.k) {  // warp-uniform conditions throughout
+                        tmem_ld16_async(taddr, va);
+                        tmem_wait16(va);
+#pragma unroll
+                        for (int c = 0; c < NC; c += 2) {
+                            const bool m1 = c + 1 < NC && jh + (c + 1) * 16 < p.k;
+                            if (m1) tmem_ld16_async(taddr + (c + 1) * 16, vb);
+                            chunk(va, c);
+                            if (!m1) break;
+                            tmem_wait16(vb);
+                            const bool m2 = c + 2 < NC && jh + (c + 2) * 16 < p.k;
+                            if (m2) tmem_ld16_async(taddr + (c + 2) * 16, va);
+                            chunk(vb, c + 1);
+                            if (!m2) break;
+                            tmem_wait16(va);
+                        }
+                    }
+                } else
 #pragma unroll 1
                 for (int c = 0; c < SW / 32; ++c) {
                     const int j0 = jh + c * 32;
@@ -684,101 +783,6 @@ __global__ void __launch_bounds__(tc_threads<NH>(), 1)
                                 besti = j0 + i;
                             }
                         }
-                    } else if (MODE == MODE_LVQ4) {
-                        // Eq. final:lvq in the library's fixed fp32 order:
-                        // key = fma(b_y, -2 A_x, N_y); key = fma(G_y, -2 b_x, key);
-                        // key = fma(-2 s_x, s_y P, key).  P is the nearest integer
-                        // to the e4m3 accumulator ((acc + 2^23) - 2^23, exact for
-                        // 0 <= acc < 2^22; P <= 225 d).  Two columns per packed op.
-                        float gb[4];
-                        int gi[4];
-#pragma unroll
-                        for (int g = 0; g < 4; ++g) {
-                            asm volatile("" ::: "memory");
-                            gb[g] = INFINITY;
-                            gi[g] = 0x7fffffff;
-#pragma unroll
-                            for (int i = 8 * g; i < 8 * g + 8; i += 2) {
-                                const float4 bg = reinterpret_cast<const float4 *>(rbuf)[(cc + i) >> 1];
-                                const float4 sn = reinterpret_cast<const float4 *>(rbuf)[128 + ((cc + i) >> 1)];
-                                const float2 P2 = fsub2(
-                                    fadd2(make_float2(__uint_as_float(v[i]), __uint_as_float(v[i + 1])),
-                                          make_float2(0x1p23f, 0x1p23f)),
-                                    make_float2(0x1p23f, 0x1p23f));
-                                float2 key = ffma2(make_float2(bg.x, bg.y), make_float2(a2, a2), make_float2(sn.z, sn.w));
-                                key = ffma2(make_float2(bg.z, bg.w), make_float2(rf2, rf2), key);
-                                const float2 t = fmul2(make_float2(sn.x, sn.y), P2);
-                                key = ffma2(make_float2(rpc, rpc), t, key);
-                                if (SEG && (j0 < cb || j0 + 32 > ce)) {  // columns outside the row's group
-                                    if (j0 + i < cb || j0 + i >= ce) key.x = INFINITY;
-                                    if (j0 + i + 1 < cb || j0 + i + 1 >= ce) key.y = INFINITY;
-                                }
-                                if (key.x < gb[g]) {
-                                    gb[g] = key.x;
-                                    gi[g] = j0 + i;
-                                }
-                                if (key.y < gb[g]) {
-                                    gb[g] = key.y;
-                                    gi[g] = j0 + i + 1;
-                                }
-                            }
-                        }
-#pragma unroll
-                        for (int g = 0; g < 4; ++g)
-                            if (gb[g] < fbest) {
-                                fbest = gb[g];
-                                besti = gi[g];
-                            }
-                    } else {
-                        // Eq. final:rabitq in Eq. rabitq_l2 in the library's fixed
-                        // fp32 order (u = fma(sd, 2P - sum ybar, bd pc),
-                        // est = fma(-2F, u, nx2 + ny2)).  The e4m3
-                        // accumulator carries a small non-integer error (~2^-12),
-                        // so P is its nearest integer, taken as (acc + 2^23) - 2^23
-                        // (exact for 0 <= acc < 2^22); 2P - sum ybar is exact.
-                        float gb[4];
-                        int gi[4];
-#pragma unroll
-                        for (int g = 0; g < 4; ++g) {
-                            asm volatile("" ::: "memory");
-                            gb[g] = INFINITY;
-                            gi[g] = 0x7fffffff;
-#pragma unroll
-                            for (int i = 8 * g; i < 8 * g + 8; i += 2) {
-                                const float4 bs = reinterpret_cast<const float4 *>(rbuf)[(cc + i) >> 1];
-                                const float4 qn = reinterpret_cast<const float4 *>(rbuf)[128 + ((cc + i) >> 1)];
-                                // packed pairs; every product here feeds an explicit fma
-                                // (no separate multiply-add the compiler could fuse)
-                                const float2 P2 = fsub2(
-                                    fadd2(make_float2(__uint_as_float(v[i]), __uint_as_float(v[i + 1])),
-                                          make_float2(0x1p23f, 0x1p23f)),
-                                    make_float2(0x1p23f, 0x1p23f));
-                                const float2 qv = ffma2(make_float2(2.0f, 2.0f), P2, make_float2(qn.x, qn.y));
-                                const float2 t = fmul2(make_float2(bs.x, bs.y), make_float2(rpc, rpc));
-                                const float2 u = ffma2(make_float2(bs.z, bs.w), qv, t);
-                                const float2 nn = fadd2(make_float2(rnx2, rnx2), make_float2(qn.z, qn.w));
-                                float2 est = ffma2(make_float2(rf2, rf2), u, nn);
-                                if (SEG && (j0 < cb || j0 + 32 > ce)) {  // columns outside the row's group
-                                    if (j0 + i < cb || j0 + i >= ce) est.x = INFINITY;
-                                    if (j0 + i + 1 < cb || j0 + i + 1 >= ce) est.y = INFINITY;
-                                }
-                                if (est.x < gb[g]) {
-                                    gb[g] = est.x;
-                                    gi[g] = j0 + i;
-                                }
-                                if (est.y < gb[g]) {
-                                    gb[g] = est.y;
-                                    gi[g] = j0 + i + 1;
-                                }
-                            }
-                        }
-                        // groups hold increasing column ranges: earlier group wins ties
-#pragma unroll
-                        for (int g = 0; g < 4; ++g)
-                            if (gb[g] < fbest) {
-                                fbest = gb[g];
-                                besti = gi[g];
-                            }
                     }
                 }
                 tc_fence_before();
@@ -1090,8 +1094,9 @@ __global__ void cprep_sq8_kernel(const uint8_t *__restrict__ C, int k, int kp, i
     }
 }
 
-// RBQ1 points: sign bits -> e4m3 bytes (bit 1 -> 1.0 = 0x38, bit 0 -> 0), row
-// stride dp bytes.  One thread per 32-bit code word writes 32 bytes.
+// RBQ1 points: sign bits -> e4m3 bytes 2 xbar - 1 (bit 1 -> +1.0 = 0x38, bit 0
+// -> -1.0 = 0xB8), row stride dp bytes (columns past d are never read: the
+// tensor map's width is d).  One thread per 32-bit code word writes 32 bytes.
 __global__ void screen_prep_rbq1_kernel(const uint32_t *__restrict__ codes, int64_t n, int d,
                                         int dp, uint8_t *__restrict__ xs) {
     const int W = (d + 31) >> 5;
@@ -1110,13 +1115,13 @@ __global__ void screen_prep_rbq1_kernel(const uint32_t *__restrict__ codes, int6
             for (int q = 0; q < 8; ++q) {
                 uint32_t v = 0;
 #pragma unroll
-                for (int u = 0; u < 4; ++u) v |= ((bits >> (4 * q + u)) & 1u) ? (0x38u << (8 * u)) : 0u;
+                for (int u = 0; u < 4; ++u) v |= (((bits >> (4 * q + u)) & 1u) ? 0x38u : 0xB8u) << (8 * u);
                 ow[q] = v;
             }
             reinterpret_cast<uint4 *>(dst)[0] = o[0];
             reinterpret_cast<uint4 *>(dst)[1] = o[1];
         } else {
-            for (int u = 0; u < nb; ++u) dst[u] = ((bits >> u) & 1u) ? 0x38 : 0x00;
+            for (int u = 0; u < nb; ++u) dst[u] = ((bits >> u) & 1u) ? 0x38 : 0xB8;
         }
     }
 }

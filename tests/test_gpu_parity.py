@@ -889,3 +889,29 @@ def test_prune_fit_sq8_trajectory_bitexact(skm):
     np.testing.assert_array_equal(a.cpu().numpy(), ao)
     np.testing.assert_array_equal(C.cpu().numpy(), Co)
     assert 0 < st["prune_complete"] <= st["prune_first_block"] <= (iters + 1) * n * k
+
+
+@pytest.mark.parametrize("d", [1024, 1000])
+def test_assign_rbq1_extreme_code_sums_exact(skm, d):
+    """The tensor path takes 2P - sum ybar straight from the e4m3 accumulator
+    (points as +-1): rows whose bits are all 1 or all 0 against centroids whose
+    SQ4 codes are almost all 15 push it to +-15 d; the estimates must still
+    equal the oracle's bit for bit."""
+    rng = np.random.default_rng(d + 1)
+    n, k = 512, 256
+    X = rng.standard_normal((n, d)).astype(np.float32)
+    X[: n // 3] = np.abs(X[: n // 3]) + 0.5  # all residuals > 0 once centred on m = 0
+    X[n // 3: 2 * n // 3] = -np.abs(X[n // 3: 2 * n // 3]) - 0.5  # all <= 0
+    m = torch.zeros(d, dtype=torch.float32, device=DEV)
+    r = skm.skm_quantize(skm.REPR_RBQ1, torch.from_numpy(X).to(DEV), fit=False, m=m)
+    pts = skm.rbq1_points(r, d)
+    h = _rbq1_host(r)
+    C = np.full((k, d), 2.0, np.float32)
+    C[np.arange(k), rng.integers(0, d, k)] = -1.0  # one code 0, the rest 15
+    C[k // 2:] += rng.integers(0, 2, (k - k // 2, d)).astype(np.float32) * 0.2
+    a, est = skm.skm_assign(pts, torch.from_numpy(C).to(DEV))
+    prep = oracle.rbq1_centroid_sq4(C, h["m"])
+    assert prep[0].mean() > 12.0
+    ao, esto = oracle.rbq1_assign(h["codes"], h["nx2"], h["F"], h["popx"], d, prep)
+    np.testing.assert_array_equal(a.cpu().numpy(), ao)
+    np.testing.assert_array_equal(est.cpu().numpy(), esto)
