@@ -464,7 +464,9 @@ int or_rbq1_exponent(const float *F, int64_t n) {
  * averaged.  F enters as the integer Fq = round(F 2^e), so the sum over the
  * members is exact and independent of order:
  *   T_i = sum Fq xbar_i,  U = sum Fq,  sum F (2 xbar_i - 1) = (2 T_i - U) 2^-e
- *   c_i = m_i + ((2 T_i - U) 2^-e / count) / sqrt(d)     (fp64, then fp32)
+ *   c_i = m_i + (2 T_i - U) * f,  f = (2^-e / sqrt(d)) / count   (fp64, then fp32)
+ * (one fp64 factor per cluster: 1/sqrt(d) rounded once, scaled by 2^-e exactly,
+ * divided by the count; the paper fixes no evaluation order).
  * Empty clusters keep their centroid.  Pinned against the fp64 mean of
  * decoded vectors (relative 1e-9) and the exact-reconstruction case. */
 void or_rbq1_update(const uint32_t *codes, const float *F, int64_t n, int d,
@@ -486,12 +488,10 @@ void or_rbq1_update(const uint32_t *codes, const float *F, int64_t n, int d,
     }
     for (int j = 0; j < k; ++j) {
         if (counts[j] == 0) continue;
+        const double f = ldexp(isd, -e) / (double)counts[j];
         for (int i = 0; i < d; ++i) {
-            double v = (double)(2 * T[(int64_t)j * d + i] - U[j]);
-            v = ldexp(v, -e);
-            v = v / (double)counts[j];
-            v = v * isd;
-            C_inout[(int64_t)j * d + i] = (float)((double)m[i] + v);
+            const double v = (double)(2 * T[(int64_t)j * d + i] - U[j]);
+            C_inout[(int64_t)j * d + i] = (float)((double)m[i] + v * f);
         }
     }
     free(T);
@@ -777,7 +777,7 @@ int or_lvq4_exponent(const float *fac, int64_t n) {
  * the integers Sq = round(s 2^e) and Bq = round(b 2^e), so the sums are exact
  * and independent of order:
  *   T_i = sum Sq xbar_i,  U = sum Bq
- *   c_i = ((T_i + U) 2^-e) / count        (int64 -> fp64, then fp32)
+ *   c_i = (T_i + U) * f,  f = 2^-e / count    (int64 -> fp64, then fp32)
  * Empty clusters keep their centroid.  Pinned against the fp64 mean of the
  * decoded members (relative 1e-8) and exactly representable members. */
 void or_lvq4_update(const uint8_t *xc, const float *xfac, int64_t n, int d, int e,
@@ -795,11 +795,10 @@ void or_lvq4_update(const uint8_t *xc, const float *xfac, int64_t n, int d, int 
     }
     for (int j = 0; j < k; ++j) {
         if (counts[j] == 0) continue;
+        const double f = ldexp(1.0, -e) / (double)counts[j];
         for (int i = 0; i < d; ++i) {
-            double v = (double)(T[(int64_t)j * d + i] + U[j]);
-            v = ldexp(v, -e);
-            v = v / (double)counts[j];
-            C_inout[(int64_t)j * d + i] = (float)v;
+            const double v = (double)(T[(int64_t)j * d + i] + U[j]);
+            C_inout[(int64_t)j * d + i] = (float)(v * f);
         }
     }
     free(T);
