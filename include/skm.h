@@ -330,12 +330,12 @@ int skm_assign_segmented(const skm_data *x, const void *C, int k, const int32_t 
  *  their centroid.  counts int64[k] (device, output).
  *   F32/BF16  c_j = mean of members (fp32 sums per cluster)
  *   SQ8       cbar_j = round-half-even(sum of member codes / count), exact
- *   RBQ1      fused decode-average: c_ji = m_i + ((2 T_ji - U_j) 2^-e
- *             / count_j) / sqrt(d) in fp64, rounded to fp32, where
+ *   RBQ1      fused decode-average: c_ji = m_i + (2 T_ji - U_j) f_j in fp64,
+ *             rounded to fp32, with f_j = (fl(1/sqrt(d)) 2^-e) / count_j, where
  *             T_ji = sum Fq xbar_i, U_j = sum Fq, Fq = round(F 2^e) (int64,
  *             exact), e = x->rbq1_exp.
- *   LVQ4      fused decode-average (Section 3.1 "LVQ4"): c_ji = ((T_ji +
- *             U_j) 2^-e) / count_j in fp64, rounded to fp32, where
+ *   LVQ4      fused decode-average (Section 3.1 "LVQ4"): c_ji = (T_ji +
+ *             U_j) f_j in fp64, rounded to fp32, f_j = 2^-e / count_j, where
  *             T_ji = sum Sq xbar_i, U_j = sum Bq, Sq = round(s 2^e),
  *             Bq = round(b 2^e) (int64, exact), e = x->rbq1_exp.
  *  Assignments outside [0, k) are skipped (not counted, not summed).

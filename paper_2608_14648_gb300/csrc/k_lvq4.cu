@@ -12,7 +12,8 @@
 //   update   fixed-point weights Sq = round(s 2^e), Bq = round(b 2^e) in the
 //            cluster-sorted order; the sums T = sum Sq xbar, U = sum Bq are
 //            exact int64 (streamed in k_ringsum.cu, or the chunk kernel here),
-//            then c = ((T + U) 2^-e) / count in fp64
+//            then c = (T + U) f in fp64 with one factor f = 2^-e / count per
+//            cluster
 //
 // Every float step that decides a code or a key is an explicit IEEE operation
 // (no contraction), in the order the oracle takes it.
@@ -327,17 +328,20 @@ __global__ void chunk_sum_lvq4_kernel(const uint32_t *__restrict__ codes, const 
     }
 }
 
+// c_i = (T_i + U) f, f = 2^-e / count formed once per cluster (one block each).
 __global__ void finalize_lvq4_kernel(const int64_t *__restrict__ partial, const int64_t *__restrict__ counts, int k,
                                      int d, int e, float *__restrict__ C) {
-    const int64_t t = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
-    if (t >= (int64_t)k * d) return;
-    const int j = (int)(t / d), i = (int)(t - (int64_t)j * d);
+    __shared__ double fs;
+    const int j = blockIdx.x;
     const int64_t c = counts[j];
-    if (c <= 0) return;
-    double v = __ll2double_rn(partial[(int64_t)j * (d + 1) + i] + partial[(int64_t)j * (d + 1) + d]);
-    v = __dmul_rn(v, ldexp(1.0, -e));
-    v = __ddiv_rn(v, (double)c);
-    C[t] = __double2float_rn(v);
+    if (c <= 0) return;  // block-uniform
+    if (threadIdx.x == 0) fs = __ddiv_rn(ldexp(1.0, -e), (double)c);
+    __syncthreads();
+    const double f = fs;
+    const int64_t *T = partial + (int64_t)j * (d + 1);
+    const int64_t U = T[d];
+    for (int i = threadIdx.x; i < d; i += blockDim.x)
+        C[(int64_t)j * d + i] = __double2float_rn(__dmul_rn(__ll2double_rn(T[i] + U), f));
 }
 
 // Forgy initial centroids: the decode-average of one member each.
@@ -356,13 +360,10 @@ __global__ void lvq4_decode_rows_kernel(const uint32_t *__restrict__ codes, cons
     const float4 f = fac[p];
     const int64_t sq = __double2ll_rn(__dmul_rn((double)f.x, pow2));
     const int64_t bq = __double2ll_rn(__dmul_rn((double)f.y, pow2));
-    const double pow2m = ldexp(1.0, -e);
+    const double g = ldexp(1.0, -e);  // the update's factor for a cluster of one member
     for (int i = threadIdx.x; i < d; i += blockDim.x) {
         const int64_t x = (codes[p * W + (i >> 3)] >> (4 * (i & 7))) & 15u;
-        double v = __ll2double_rn(sq * x + bq);
-        v = __dmul_rn(v, pow2m);
-        v = __ddiv_rn(v, 1.0);
-        out[(int64_t)j * d + i] = __double2float_rn(v);
+        out[(int64_t)j * d + i] = __double2float_rn(__dmul_rn(__ll2double_rn(sq * x + bq), g));
     }
 }
 
@@ -435,8 +436,7 @@ cudaError_t launch_chunk_sum_lvq4(const uint32_t *codes, const uint32_t *sq, con
 
 cudaError_t launch_finalize_lvq4(const int64_t *partial, const int64_t *counts, int k, int d, int e, float *C_inout,
                                  cudaStream_t st) {
-    const int64_t tot = (int64_t)k * d;
-    finalize_lvq4_kernel<<<(unsigned)((tot + 255) / 256), 256, 0, st>>>(partial, counts, k, d, e, C_inout);
+    finalize_lvq4_kernel<<<k, 256, 0, st>>>(partial, counts, k, d, e, C_inout);
     return launched();
 }
 

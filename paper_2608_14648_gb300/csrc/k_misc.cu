@@ -45,14 +45,11 @@ __global__ void rbq1_decode_rows_kernel(const uint32_t *__restrict__ codes,
         return;
     }
     const int64_t fq = __double2ll_rn(__dmul_rn((double)F[p], ldexp(1.0, e)));
-    const double pow2m = ldexp(1.0, -e);
-    const double isd = __ddiv_rn(1.0, __dsqrt_rn((double)d));
+    // the update's factor for a cluster of one member: fl(1/sqrt(d)) 2^-e
+    const double f = __dmul_rn(__ddiv_rn(1.0, __dsqrt_rn((double)d)), ldexp(1.0, -e));
     for (int i = threadIdx.x; i < d; i += blockDim.x) {
         const int64_t T = ((codes[p * W + (i >> 5)] >> (i & 31)) & 1u) ? fq : 0;
-        double v = __ll2double_rn(2 * T - fq);
-        v = __dmul_rn(v, pow2m);
-        v = __ddiv_rn(v, 1.0);
-        v = __dmul_rn(v, isd);
+        const double v = __dmul_rn(__ll2double_rn(2 * T - fq), f);
         out[(int64_t)j * d + i] = __double2float_rn(__dadd_rn((double)m[i], v));
     }
 }

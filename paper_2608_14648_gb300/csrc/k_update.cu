@@ -278,14 +278,10 @@ cudaError_t launch_segsum_sq8(const uint8_t *X, int d, const int32_t *perm,
 // ------------------------------------------------------ segmented sums: RBQ1
 // Fused decode-average with exact fixed-point sums: Fq = rint(F 2^e),
 // T_i = sum Fq xbar_i, U = sum Fq;
-// c_i = m_i + (((2 T_i - U) 2^-e) / count) / sqrt(d) in fp64 -> fp32.
-__device__ __forceinline__ float rbq1_finish(int64_t T, int64_t U, int64_t cnt, float m,
-                                             double pow2m, double isd) {
-    double v = __ll2double_rn(2 * T - U);
-    v = __dmul_rn(v, pow2m);
-    v = __ddiv_rn(v, (double)cnt);
-    v = __dmul_rn(v, isd);
-    return __double2float_rn(__dadd_rn((double)m, v));
+// c_i = m_i + (2 T_i - U) f in fp64 -> fp32, with one factor per cluster
+// f = (fl(1/sqrt(d)) 2^-e) / count.
+__device__ __forceinline__ float rbq1_finish(int64_t T, int64_t U, float m, double f) {
+    return __double2float_rn(__dadd_rn((double)m, __dmul_rn(__ll2double_rn(2 * T - U), f)));
 }
 
 // Fixed-point weights Fq = rint(F 2^e), once per update call, written in the
@@ -573,25 +569,30 @@ cudaError_t launch_finalize_sq8(const int64_t *partial, const int64_t *counts, i
     return launched();
 }
 
+// One block per cluster: the factor f (one fp64 square root and division) is
+// formed once and shared; GB300's fp64 rate makes per-element divisions the
+// cost of this step otherwise.
 __global__ void finalize_rbq1_kernel(const int64_t *__restrict__ partial,
                                      const int64_t *__restrict__ counts, int k, int d,
                                      const float *__restrict__ m, int e, float *__restrict__ C) {
-    const int64_t t = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
-    if (t >= (int64_t)k * d) return;
-    const int j = (int)(t / d), i = (int)(t - (int64_t)j * d);
+    __shared__ double fs;
+    const int j = blockIdx.x;
     const int64_t c = counts[j];
-    if (c <= 0) return;
-    const double pow2m = ldexp(1.0, -e);
-    const double isd = __ddiv_rn(1.0, __dsqrt_rn((double)d));
-    C[t] = rbq1_finish(partial[(int64_t)j * (d + 1) + i], partial[(int64_t)j * (d + 1) + d], c,
-                       m[i], pow2m, isd);
+    if (c <= 0) return;  // block-uniform
+    if (threadIdx.x == 0) {
+        const double isd = __ddiv_rn(1.0, __dsqrt_rn((double)d));
+        fs = __ddiv_rn(__dmul_rn(isd, ldexp(1.0, -e)), (double)c);
+    }
+    __syncthreads();
+    const double f = fs;
+    const int64_t *T = partial + (int64_t)j * (d + 1);
+    const int64_t U = T[d];
+    for (int i = threadIdx.x; i < d; i += blockDim.x) C[(int64_t)j * d + i] = rbq1_finish(T[i], U, m[i], f);
 }
 
 cudaError_t launch_finalize_rbq1(const int64_t *partial, const int64_t *counts, int k, int d,
                                  const float *m, int e, float *C_inout, cudaStream_t st) {
-    const int64_t tot = (int64_t)k * d;
-    finalize_rbq1_kernel<<<(unsigned)((tot + 255) / 256), 256, 0, st>>>(partial, counts, k, d, m,
-                                                                        e, C_inout);
+    finalize_rbq1_kernel<<<k, 256, 0, st>>>(partial, counts, k, d, m, e, C_inout);
     return launched();
 }
 
