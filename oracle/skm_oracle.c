@@ -446,8 +446,9 @@ void or_rbq1_assign(const uint32_t *codes, const float *nx2, const float *F,
     }
 }
 
-/* Fixed-point exponent for the decode-average: e = 37 - ceil(log2 max F),
- * so F * 2^e <= 2^37; e = 0 when every F is 0. */
+/* Fixed-point exponent for the decode-average: e = 24 - ceil(log2 max F),
+ * so F * 2^e <= 2^24 (the largest F keeps its 24-bit fp32 precision) and
+ * sums over up to 2^24 members stay exact in int64; e = 0 when every F is 0. */
 int or_rbq1_exponent(const float *F, int64_t n) {
     float mx = 0.0f;
     for (int64_t p = 0; p < n; ++p)
@@ -456,7 +457,7 @@ int or_rbq1_exponent(const float *F, int64_t n) {
     int ex;
     double fr = frexp((double)mx, &ex); /* mx = fr * 2^ex, fr in [0.5, 1) */
     int c = (fr == 0.5) ? ex - 1 : ex;  /* ceil(log2 mx) */
-    return 37 - c;
+    return 24 - c;
 }
 
 /* Fused decode-average (Section 3.1 "RabitQ", last paragraph): the member
