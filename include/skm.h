@@ -219,8 +219,9 @@ typedef struct skm_quant_params {
 int skm_quantize(int repr, const float *X, int64_t n, int d, skm_quant_params *qp,
                  void *codes, void *ws, size_t ws_bytes, void *stream);
 
-/* Fixed-point exponent e of the RBQ1 decode-average: e = 37 - ceil(log2 max F)
- * (0 when every F is 0), so round(F 2^e) <= 2^37 and the per-cluster sums of
+/* Fixed-point exponent e of the RBQ1 decode-average: e = 24 - ceil(log2 max F)
+ * (0 when every F is 0), so round(F 2^e) <= 2^24 (the largest F keeps its
+ * 24-bit precision) and the per-cluster sums of
  * up to 2^24 points are exact in int64.  Writes *e_host; synchronises. */
 int skm_rbq1_exponent(const float *F, int64_t n, int *e_host, void *ws, size_t ws_bytes,
                       void *stream);

@@ -267,7 +267,7 @@ cudaError_t launch_rbq1_encode(const float *X, int64_t n, int d, const float *m,
 }
 
 // max F (F >= 0, so the IEEE bit pattern orders like an unsigned integer),
-// then e = 37 - ceil(log2 max F), e = 0 when max F == 0.
+// then e = 24 - ceil(log2 max F), e = 0 when max F == 0.
 __global__ void rbq1_maxbits_kernel(const float *__restrict__ F, int64_t n,
                                     unsigned int *__restrict__ maxbits) {
     unsigned int mx = 0;
@@ -290,7 +290,7 @@ __global__ void rbq1_exponent_kernel(const unsigned int *__restrict__ maxbits, i
     int ex;
     const double fr = frexp((double)mx, &ex);
     const int c = (fr == 0.5) ? ex - 1 : ex;
-    *e = 37 - c;
+    *e = 24 - c;
 }
 
 cudaError_t launch_rbq1_exponent(const float *F, int64_t n, unsigned int *maxbits, int *e_dev,

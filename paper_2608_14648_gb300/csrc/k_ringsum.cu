@@ -314,16 +314,16 @@ __global__ void __launch_bounds__(RS_THREADS) ring_sum_float_kernel(
 // ------------------------------------------------------------- 1-bit rows
 // T[c][i] += Fq for every member with bit i set; T[c][d] += Fq (= U).
 // Lane l holds dimension l of each of the W = 4 W4 code words.  Inside a run
-// (at most RS_ROWS rows between flushes) Fq = hi 2^20 + lo is accumulated as
-// two 32-bit sums, which cannot overflow (Fq <= 2^37: sum lo < 2^27, sum hi
-// <= 2^24), so each (row, dimension) costs one test and two predicated adds.
+// (at most RS_ROWS = 128 rows between flushes) the sums fit 32 bits
+// (Fq <= 2^24), so each (row, dimension) costs one bit test and one
+// predicated add.
 template <int W4>
 struct Rbq1Cons {
     const int32_t *scl;
     const int64_t *fqs;  // Fq in sorted order
     unsigned long long *T;
     int d;
-    uint32_t alo[4 * W4], ahi[4 * W4];
+    uint32_t acc[4 * W4];
     int64_t usum;
     int cur;
     int64_t q0;
@@ -334,10 +334,8 @@ struct Rbq1Cons {
 #pragma unroll
         for (int t = 0; t < 4 * W4; ++t) {
             const int col = 32 * t + lane;
-            const unsigned long long v = ((unsigned long long)ahi[t] << 20) + alo[t];
-            if (col < d && v) atomicAdd(T + (int64_t)c * (d + 1) + col, v);
-            alo[t] = 0;
-            ahi[t] = 0;
+            if (col < d && acc[t]) atomicAdd(T + (int64_t)c * (d + 1) + col, (unsigned long long)acc[t]);
+            acc[t] = 0;
         }
         if (lane == 0 && usum) atomicAdd(T + (int64_t)c * (d + 1) + d, (unsigned long long)usum);
         usum = 0;
@@ -346,10 +344,7 @@ struct Rbq1Cons {
         q0 = q0_;
         cnt = cnt_;
 #pragma unroll
-        for (int t = 0; t < 4 * W4; ++t) {
-            alo[t] = 0;
-            ahi[t] = 0;
-        }
+        for (int t = 0; t < 4 * W4; ++t) acc[t] = 0;
         usum = 0;
         clw = lane < cnt ? __ldg(scl + q0 + lane) : -1;
         cln = 32 + lane < cnt ? __ldg(scl + q0 + 32 + lane) : -1;
@@ -372,16 +367,16 @@ struct Rbq1Cons {
             cur = c;
         }
         usum += fq;
-        const uint32_t flo = (uint32_t)fq & 0xfffffu, fhi = (uint32_t)(fq >> 20);
+        const uint32_t f32 = (uint32_t)fq;
         const uint32_t lm = 1u << lane;
         const uint4 *w4 = reinterpret_cast<const uint4 *>(slot);
 #pragma unroll
         for (int g = 0; g < W4; ++g) {
             const uint4 wv = w4[g];  // broadcast: every lane reads the same 16 bytes
-            add_if_bit2(alo[4 * g + 0], ahi[4 * g + 0], wv.x, lm, flo, fhi);
-            add_if_bit2(alo[4 * g + 1], ahi[4 * g + 1], wv.y, lm, flo, fhi);
-            add_if_bit2(alo[4 * g + 2], ahi[4 * g + 2], wv.z, lm, flo, fhi);
-            add_if_bit2(alo[4 * g + 3], ahi[4 * g + 3], wv.w, lm, flo, fhi);
+            add_if_bit(acc[4 * g + 0], wv.x, lm, f32);
+            add_if_bit(acc[4 * g + 1], wv.y, lm, f32);
+            add_if_bit(acc[4 * g + 2], wv.z, lm, f32);
+            add_if_bit(acc[4 * g + 3], wv.w, lm, f32);
         }
     }
     __device__ __forceinline__ void finish(int lane) { flush(cur, lane); }

@@ -55,6 +55,17 @@ struct Carver {
 inline int words_of(int d) { return (d + 31) / 32; }
 inline int64_t cdiv(int64_t a, int64_t b) { return (a + b - 1) / b; }
 
+// acc += f when (word & mask) != 0: one bit test and one predicated 32-bit add
+// (the 1-bit decode-average sums of a run of rows).
+__device__ __forceinline__ void add_if_bit(uint32_t &acc, uint32_t word, uint32_t mask, uint32_t f) {
+    asm("{\n\t.reg .pred p;\n\t"
+        "and.b32 %1, %1, %2;\n\t"
+        "setp.ne.u32 p, %1, 0;\n\t"
+        "@p add.u32 %0, %0, %3;\n\t}"
+        : "+r"(acc), "+r"(word)
+        : "r"(mask), "r"(f));
+}
+
 // (lo, hi) += (flo, fhi) when (word & mask) != 0, as two predicated 32-bit
 // adds (no branch, no carry); used by the 1-bit decode-average sums, which
 // split each fixed-point weight as hi 2^20 + lo.
