@@ -78,6 +78,8 @@ def lib():
                 "or_rbq1_centroid_sq4": ([vp, i32, i32, vp, vp, vp, vp, vp, vp], None),
                 "or_rbq1_assign": ([vp, vp, vp, vp, i64, i32, vp, vp, vp, vp, vp, i32, vp, vp], None),
                 "or_rbq1_exponent": ([vp, i64], i32),
+                "or_rbq1_centroid_sym": ([vp, i32, i32, vp, vp, vp, vp], None),
+                "or_rbq1_assign_sym": ([vp, vp, vp, i64, i32, vp, vp, vp, i32, vp, vp], None),
                 "or_rbq1_update": ([vp, vp, i64, i32, vp, i32, vp, i32, vp, vp], None),
                 "or_project": ([vp, i64, i32, vp, vp, i32, vp], None),
                 "or_mean_cov": ([vp, i64, i32, vp, vp], None),
@@ -300,6 +302,44 @@ def rbq1_assign(codes, nx2, F, popx, d, prep):
         _p(_c(ny2, np.float32)), k, _p(a), _p(est),
     )
     return a, est
+
+
+def rbq1_centroid_sym(C, m):
+    """Symmetric 1-bit centroid side: (bits uint32[k, W], fy f32[k], ny2 f32[k])."""
+    C = _c(C, np.float32)
+    k, d = C.shape
+    W = (d + 31) // 32
+    yb = np.empty((k, W), np.uint32)
+    fy = np.empty(k, np.float32)
+    ny2 = np.empty(k, np.float32)
+    lib().or_rbq1_centroid_sym(_p(C), k, d, _p(_c(m, np.float32)), _p(yb), _p(fy), _p(ny2))
+    return yb, fy, ny2
+
+
+def rbq1_assign_sym(codes, nx2, F, d, prep):
+    """XOR + POPCOUNT estimate against binarized centroids; (assign, est)."""
+    codes = _c(codes, np.uint32)
+    n = codes.shape[0]
+    yb, fy, ny2 = prep
+    k = yb.shape[0]
+    a = np.empty(n, np.int32)
+    est = np.empty(n, np.float32)
+    lib().or_rbq1_assign_sym(_p(codes), _p(_c(nx2, np.float32)), _p(_c(F, np.float32)), n, d, _p(_c(yb, np.uint32)),
+                             _p(_c(fy, np.float32)), _p(_c(ny2, np.float32)), k, _p(a), _p(est))
+    return a, est
+
+
+def lloyd_rbq1_sym(codes, nx2, F, popx, d, m, C0, iters, e=None):
+    """Lloyd with the symmetric estimate in the assignment (the update is the
+    fused decode-average of the points, as in the asymmetric variant)."""
+    if e is None:
+        e = rbq1_exponent(F)
+    C = np.array(C0, np.float32, copy=True)
+    for _ in range(iters):
+        a, _ = rbq1_assign_sym(codes, nx2, F, d, rbq1_centroid_sym(C, m))
+        C, _ = rbq1_update(codes, F, d, m, e, a, C)
+    a, _ = rbq1_assign_sym(codes, nx2, F, d, rbq1_centroid_sym(C, m))
+    return C, a
 
 
 def rbq1_exponent(F) -> int:

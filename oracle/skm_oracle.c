@@ -446,6 +446,76 @@ void or_rbq1_assign(const uint32_t *codes, const float *nx2, const float *F,
     }
 }
 
+/* Symmetric 1-bit variant (the centroid binarized like a point; XOR +
+ * POPCOUNT).  Applying RabitQ's estimate <o, q> ~ <obar, q> / <obar, o> to
+ * both unit vectors gives <x - m, y - m> ~ F_x F_y <obar_x, obar_y> with
+ * obar = (2 bit - 1) / sqrt(d), i.e. F_x F_y (d - 2 h) / d for the Hamming
+ * distance h = popc(xbar XOR ybar).  Centroid side, once per assignment:
+ * rho = c - m (fp32), bits (rho_i > 0), ny2 = ||rho||^2 in the blocked fp64
+ * order, l1 = ||rho||_1 in the same blocked order, and
+ *   fy = fl32((ny2 / l1) / sqrt(d))   (fp64; fy = 0 when l1 = 0)  = F_y / d.
+ * Estimate, fp32, in this order: u = fy * (float)(d - 2h) (exact integer),
+ * est = fma(-2 F_x, u, nx2 + ny2); argmin, ties to the lowest index. */
+static double sumabs_blocked(const float *r, int d) {
+    double q = 0.0;
+    for (int w = 0; w < (d + 31) / 32; ++w) {
+        double v[32];
+        for (int l = 0; l < 32; ++l) {
+            int i = 32 * w + l;
+            v[l] = (i < d) ? fabs((double)r[i]) : 0.0;
+        }
+        for (int o = 16; o >= 1; o >>= 1)
+            for (int l = 0; l < o; ++l) v[l] = v[l] + v[l + o];
+        q = q + v[0];
+    }
+    return q;
+}
+
+void or_rbq1_centroid_sym(const float *C, int k, int d, const float *m, uint32_t *ybits, float *fy,
+                          float *ny2) {
+    const int W = (d + 31) / 32;
+    float *rho = (float *)malloc(sizeof(float) * (size_t)d);
+    for (int j = 0; j < k; ++j) {
+        uint32_t *yw = ybits + (int64_t)j * W;
+        for (int w = 0; w < W; ++w) yw[w] = 0u;
+        for (int i = 0; i < d; ++i) {
+            rho[i] = C[(int64_t)j * d + i] - m[i];
+            if (rho[i] > 0.0f) yw[i / 32] |= 1u << (i % 32);
+        }
+        const double q2 = sumsq_blocked(rho, d);
+        const double l1 = sumabs_blocked(rho, d);
+        ny2[j] = (float)q2;
+        fy[j] = (l1 > 0.0) ? (float)((q2 / l1) / sqrt((double)d)) : 0.0f;
+    }
+    free(rho);
+}
+
+void or_rbq1_assign_sym(const uint32_t *codes, const float *nx2, const float *F, int64_t n, int d,
+                        const uint32_t *ybits, const float *fy, const float *ny2, int k, int32_t *assign,
+                        float *est_best) {
+    const int W = (d + 31) / 32;
+#pragma omp parallel for schedule(dynamic, 16)
+    for (int64_t p = 0; p < n; ++p) {
+        const uint32_t *cw = codes + p * (int64_t)W;
+        const float f2 = -2.0f * F[p];
+        float best = INFINITY;
+        int32_t a = -1;
+        for (int j = 0; j < k; ++j) {
+            int h = 0; /* Hamming distance, bit by bit */
+            for (int i = 0; i < d; ++i)
+                h += (int)(((cw[i / 32] ^ ybits[(int64_t)j * W + i / 32]) >> (i % 32)) & 1u);
+            const float u = fy[j] * (float)(d - 2 * h);
+            const float est = fmaf(f2, u, nx2[p] + ny2[j]);
+            if (est < best) {
+                best = est;
+                a = j;
+            }
+        }
+        assign[p] = a;
+        if (est_best) est_best[p] = best;
+    }
+}
+
 /* Fixed-point exponent for the decode-average: e = 24 - ceil(log2 max F),
  * so F * 2^e <= 2^24 (the largest F keeps its 24-bit fp32 precision) and
  * sums over up to 2^24 members stay exact in int64; e = 0 when every F is 0. */

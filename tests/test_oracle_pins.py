@@ -713,3 +713,46 @@ def test_hierarchical_lvq4_one_meso_cluster_equals_lloyd():
     C2, a2 = oracle.lloyd_lvq4(codes, fac, oracle.lvq4_decode_points(codes, fac, e, init), 3, e=e)
     np.testing.assert_array_equal(C, C2)
     np.testing.assert_array_equal(a, a2)
+
+
+# ------------------------------------------------- symmetric 1-bit (XOR + POPCOUNT)
+def test_rbq1_symmetric_estimate_matches_formula_and_hamming():
+    """Estimate = nx2 + ny2 - 2 F_x F_y (d - 2 h) / d with h the Hamming
+    distance of the sign codes (numpy popcount of the XOR), in fp64."""
+    r = _rng(48)
+    n, d, k = 80, 70, 9
+    X = r.standard_normal((n, d)).astype(np.float32)
+    C = r.standard_normal((k, d)).astype(np.float32)
+    m = oracle.rbq1_mean(X)
+    codes, nx2, F, popx = oracle.rbq1_encode(X, m)
+    yb, fy, ny2 = oracle.rbq1_centroid_sym(C, m)
+    # the centroid side is the point encoder's sign code and factor
+    cc, cn2, cF, _ = oracle.rbq1_encode(C, m)
+    np.testing.assert_array_equal(yb, cc)
+    np.testing.assert_allclose(ny2, cn2, rtol=1e-6)
+    np.testing.assert_allclose(fy * d, cF, rtol=1e-5)
+    a, est = oracle.rbq1_assign_sym(codes, nx2, F, d, (yb, fy, ny2))
+    bx = np.unpackbits(codes.view(np.uint8), axis=1, bitorder="little")[:, :d].astype(np.int64)
+    by = np.unpackbits(yb.view(np.uint8), axis=1, bitorder="little")[:, :d].astype(np.int64)
+    h = (bx[:, None, :] != by[None, :, :]).sum(-1)
+    E = nx2[:, None].astype(np.float64) + ny2[None, :] - 2.0 * F[:, None] * cF[None, :] * (d - 2 * h) / d
+    np.testing.assert_allclose(est, E[np.arange(n), a], rtol=2e-5, atol=1e-4)
+    srt = np.sort(E, 1)
+    clear = (srt[:, 1] - srt[:, 0]) > 1e-4 * np.abs(srt).max()
+    np.testing.assert_array_equal(a[clear], E.argmin(1)[clear])
+
+
+def test_rbq1_symmetric_exact_for_sign_constant_vectors():
+    """Residuals of constant magnitude are reconstructed exactly by
+    F (2 bit - 1) / sqrt(d), so the symmetric estimate is the true squared
+    distance (up to rounding)."""
+    r = _rng(49)
+    n, k, d = 20, 6, 64
+    m = np.zeros(d, np.float32)
+    X = (r.choice([-1.0, 1.0], (n, d)) * r.uniform(0.5, 2.0, (n, 1))).astype(np.float32)
+    C = (r.choice([-1.0, 1.0], (k, d)) * r.uniform(0.5, 2.0, (k, 1))).astype(np.float32)
+    codes, nx2, F, _ = oracle.rbq1_encode(X, m)
+    a, est = oracle.rbq1_assign_sym(codes, nx2, F, d, oracle.rbq1_centroid_sym(C, m))
+    D = cdist(X.astype(np.float64), C.astype(np.float64), "sqeuclidean")
+    np.testing.assert_allclose(est, D[np.arange(n), a], rtol=1e-5)
+    np.testing.assert_array_equal(a, D.argmin(1))
