@@ -597,6 +597,9 @@ def run_config(args):
         pR = skm.rbq1_points(q, spec.d).with_screen()
         CR, _, _, _, _ = skm.skm_fit(pR, k, 0, init_idx=idx, want_objective=False, want_dist=False)
         runs.append(("rbq1", pR, CR, spec.d, 2 * bf16_peak, "e4m3"))
+        if args.symmetric:
+            runs.append(("rbq1_symmetric", pR.with_flags(skm.FLAG_SYMMETRIC), CR.clone(), spec.d, 2 * bf16_peak,
+                         "e4m3"))
     if args.config in ("c1", "c2"):
         pL = skm.lvq4_points(skm.skm_quantize(skm.REPR_LVQ4, X), spec.d).with_screen()
         CL, _, _, _, _ = skm.skm_fit(pL, k, 0, init_idx=idx, want_objective=False, want_dist=False)
@@ -698,6 +701,8 @@ def main():
     ap.add_argument("--iters", type=int, default=10)
     ap.add_argument("--lvq4", action="store_true", help="with --config c3: also time LVQ4 on the rotated points")
     ap.add_argument("--prune", action="store_true", help="with --config c2: also time SQ8 with exact pruning")
+    ap.add_argument("--symmetric", action="store_true",
+                    help="with --config c1: also time the symmetric 1-bit assignment (binarized centroids)")
     ap.add_argument("--hier", action="store_true",
                     help="with --config: flat Lloyd fit against hierarchical k-means (m = sqrt k)")
     args = ap.parse_args()

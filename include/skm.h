@@ -72,7 +72,17 @@ enum {
      * current best) instead of the tensor-core path.  Same result (the fp32
      * nearest centroid; for SQ8 the exact integer code-space nearest, with
      * integer partial sums). */
-    SKM_FLAG_PRUNE = 1
+    SKM_FLAG_PRUNE = 1,
+    /* RBQ1 only: symmetric 1-bit assignment -- every centroid is binarized
+     * like a point (rho = c - m, bit = rho_i > 0) instead of SQ4-coded, and
+     * the estimate of Eq. rabitq_l2 uses RabitQ's <o, q> ~ <obar, q>/<obar, o>
+     * on both sides: <x - m, c - m> ~ F_x F_y (d - 2 h) / d with h the Hamming
+     * distance (XOR + POPCOUNT) of the sign codes.  fp32 order: fy =
+     * fl32((||rho||^2 / ||rho||_1) / sqrt(d)) per centroid (fp64, blocked
+     * order), u = fy (d - 2 h), est = fma(-2 F, u, nx2 + ||rho||^2).  Tensor
+     * cores (e4m3 +-1 codes on both sides) for d <= 1024, XOR + POPC beyond.
+     * The update is unchanged (the points' fused decode-average). */
+    SKM_FLAG_SYMMETRIC = 2
 };
 
 /* Points being clustered.  Which fields are read depends on repr. */

@@ -97,6 +97,75 @@ __global__ void __launch_bounds__(RBQ1_THREADS) assign_rbq1_kernel(
     }
 }
 
+// Symmetric variant (binarized centroids): Hamming distance h by XOR + POPC,
+// est = fma(-2 F, fy (d - 2h), nx2 + ny2) in that fp32 order.  One thread per
+// point; tiles of SYM_KT centroids' sign words in shared memory (broadcast
+// reads), the point's words from global memory (L1-resident across a tile).
+constexpr int SYM_KT = 32;
+__global__ void __launch_bounds__(RBQ1_THREADS) assign_rbq1_sym_kernel(
+    const uint32_t *__restrict__ codes, const float *__restrict__ nx2, const float *__restrict__ F, int64_t n, int d,
+    const uint32_t *__restrict__ yw, const Rbq1CInfo *__restrict__ info, int k, int32_t *__restrict__ assign,
+    float *__restrict__ dist) {
+    extern __shared__ uint32_t sy[];  // [SYM_KT][W]
+    const int W = (d + 31) >> 5;
+    const int64_t p = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
+    const bool valid = p < n;
+    const uint32_t *xr = codes + (valid ? p : 0) * W;
+    const float f2 = valid ? __fmul_rn(-2.0f, F[p]) : 0.0f;
+    const float xn = valid ? nx2[p] : 0.0f;
+    float best = INFINITY;
+    int32_t besti = 0;
+    for (int j0 = 0; j0 < k; j0 += SYM_KT) {
+        __syncthreads();
+        for (int t = threadIdx.x; t < SYM_KT * W; t += blockDim.x) {
+            const int c = t / W, w = t - c * W;
+            sy[t] = (j0 + c < k) ? yw[(int64_t)(j0 + c) * W + w] : 0u;
+        }
+        __syncthreads();
+        if (!valid) continue;
+        int h[SYM_KT];
+#pragma unroll
+        for (int c = 0; c < SYM_KT; ++c) h[c] = 0;
+        for (int w = 0; w < W; ++w) {
+            const uint32_t xw = xr[w];
+#pragma unroll
+            for (int c = 0; c < SYM_KT; ++c) h[c] += __popc(xw ^ sy[c * W + w]);
+        }
+#pragma unroll
+        for (int c = 0; c < SYM_KT; ++c) {
+            const int j = j0 + c;
+            if (j < k) {
+                const Rbq1CInfo in = info[j];
+                const float u = __fmul_rn(in.sd, __int2float_rn(d - 2 * h[c]));
+                const float est = __fmaf_rn(f2, u, __fadd_rn(xn, in.ny2));
+                if (est < best) {
+                    best = est;
+                    besti = j;
+                }
+            }
+        }
+    }
+    if (valid) {
+        assign[p] = besti;
+        if (dist) dist[p] = best;
+    }
+}
+
+cudaError_t launch_assign_rbq1_sym(const uint32_t *codes, const float *nx2, const float *F, int64_t n, int d,
+                                   const uint32_t *yw, const Rbq1CInfo *info, int k, int32_t *assign, float *dist,
+                                   cudaStream_t st) {
+    if (n == 0) return cudaSuccess;
+    const size_t smem = (size_t)SYM_KT * ((d + 31) >> 5) * sizeof(uint32_t);
+    if (smem > 48 * 1024) {
+        const cudaError_t e =
+            cudaFuncSetAttribute(assign_rbq1_sym_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+        if (e != cudaSuccess) return e;
+    }
+    assign_rbq1_sym_kernel<<<(unsigned)((n + RBQ1_THREADS - 1) / RBQ1_THREADS), RBQ1_THREADS, smem, st>>>(
+        codes, nx2, F, n, d, yw, info, k, assign, dist);
+    return launched();
+}
+
 cudaError_t launch_assign_rbq1(const uint32_t *codes, const float *nx2, const float *F,
                                const int32_t *popx, int64_t n, int d, const uint4 *planes,
                                const Rbq1CInfo *info, int k, int32_t *assign, float *dist,

@@ -58,6 +58,8 @@ extern "C" int skm_assign_rbq1_noalloc(const skm_data *x, const float *C, int k,
                                        float *dist, void *stream) {
     if (!x || x->repr != SKM_REPR_RBQ1)
         return set_error(SKM_ERR_INVALID_ARG, "skm_assign_rbq1_noalloc needs RBQ1 points");
+    if (x->flags & SKM_FLAG_SYMMETRIC)
+        return set_error(SKM_ERR_UNSUPPORTED, "skm_assign_rbq1_noalloc: the asymmetric estimate only");
     if (!x->x || !x->nx2 || !x->F || !x->popx || !x->m || !C || !assign)
         return set_error(SKM_ERR_INVALID_ARG, "NULL pointer");
     if (x->d < 1 || x->d > 4096 || x->n < 1 || x->n > (int64_t(1) << 24))

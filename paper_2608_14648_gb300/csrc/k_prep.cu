@@ -104,6 +104,55 @@ cudaError_t launch_rbq1_cprep_tc(const float *C, int k, int d, const float *m, u
     return launch_cprep_common(C, k, d, m, nullptr, info, yq, dq, st);
 }
 
+// Symmetric 1-bit variant: the centroid residual rho = c - m binarized like a
+// point (bit = rho_i > 0); ||rho||^2 and ||rho||_1 in fp64, pairwise inside
+// 32-dimension blocks, blocks in order; fy = fl32((||rho||^2 / ||rho||_1) /
+// sqrt(d)) = F_y / d (0 when rho = 0).  Outputs: e4m3 +-1 codes (yq, row
+// stride dq) and/or sign words (yw), and info = (bd 0, sd fy, sumy 0, ny2), so
+// the tensor epilogue's u = fma(sd, acc, bd pc) is fy (d - 2h).
+__global__ void __launch_bounds__(CPREP_WARPS * 32) rbq1_cprep_sym_kernel(
+    const float *__restrict__ C, int k, int d, const float *__restrict__ m, uint8_t *__restrict__ yq, int dq,
+    uint32_t *__restrict__ yw, Rbq1CInfo *__restrict__ info) {
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int j = blockIdx.x * CPREP_WARPS + warp;
+    if (j >= k) return;  // warp-uniform
+    const float *c = C + (int64_t)j * d;
+    const int W = (d + 31) >> 5;
+    double q2 = 0.0, l1 = 0.0;
+    for (int w = 0; w < W; ++w) {
+        const int i = 32 * w + lane;
+        const float r = (i < d) ? __fsub_rn(c[i], m[i]) : 0.0f;
+        double sq = (i < d) ? __dmul_rn((double)r, (double)r) : 0.0;
+        double ab = (i < d) ? fabs((double)r) : 0.0;
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) {
+            sq = __dadd_rn(sq, __shfl_xor_sync(0xffffffffu, sq, o));
+            ab = __dadd_rn(ab, __shfl_xor_sync(0xffffffffu, ab, o));
+        }
+        q2 = __dadd_rn(q2, sq);
+        l1 = __dadd_rn(l1, ab);
+        const bool bit = (i < d) && r > 0.0f;
+        if (yq && i < d) yq[(int64_t)j * dq + i] = bit ? 0x38 : 0xB8;
+        const uint32_t word = __ballot_sync(0xffffffffu, bit);
+        if (yw && lane == 0) yw[(int64_t)j * W + w] = word;
+    }
+    if (lane == 0) {
+        Rbq1CInfo in;
+        in.bd = 0.0f;
+        in.sd = (l1 > 0.0) ? __double2float_rn(__ddiv_rn(__ddiv_rn(q2, l1), __dsqrt_rn((double)d))) : 0.0f;
+        in.sumy = 0;
+        in.ny2 = __double2float_rn(q2);
+        info[j] = in;
+    }
+}
+
+cudaError_t launch_rbq1_cprep_sym(const float *C, int k, int d, const float *m, uint8_t *yq, int dq, uint32_t *yw,
+                                  Rbq1CInfo *info, cudaStream_t st) {
+    rbq1_cprep_sym_kernel<<<(k + CPREP_WARPS - 1) / CPREP_WARPS, CPREP_WARPS * 32, 0, st>>>(C, k, d, m, yq, dq, yw,
+                                                                                        info);
+    return launched();
+}
+
 // sum_i code_i^2 per row (exact, fits int32 for d <= 4096); one warp per row.
 __global__ void row_sqnorm_u8_kernel(const uint8_t *__restrict__ codes, int64_t n, int d,
                                      int32_t *__restrict__ out) {

@@ -1705,8 +1705,12 @@ int tc_assign_rbq1(const skm_data *x, const float *C, int k, int32_t *assign, fl
     }
     ScreenView v = screen_view(x->repr, n, d, x->x, screen);
     const int kp = (int)(cdiv(k, BN) * BN);
-    SKM_CUDA_TRY(launch_rbq1_cprep_tc(C, k, d, x->m, reinterpret_cast<uint8_t *>(b.cs), dp, b.rinfo,
-                                      st));
+    if (x->flags & SKM_FLAG_SYMMETRIC)
+        SKM_CUDA_TRY(launch_rbq1_cprep_sym(C, k, d, x->m, reinterpret_cast<uint8_t *>(b.cs), dp, nullptr, b.rinfo,
+                                           st));
+    else
+        SKM_CUDA_TRY(launch_rbq1_cprep_tc(C, k, d, x->m, reinterpret_cast<uint8_t *>(b.cs), dp, b.rinfo,
+                                          st));
     pack_rbq1_pairs_kernel<<<(kp / 2 + 255) / 256, 256, 0, st>>>(b.rinfo, k, kp, b.rpair_bs,
                                                                  b.rpair_qn);
     SKM_CUDA_TRY(launched());

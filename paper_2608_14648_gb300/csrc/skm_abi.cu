@@ -61,6 +61,8 @@ static int check_data(const skm_data *x, bool need_codes = true) {
         if (!x->nx2 || !x->F || !x->popx || !x->m)
             return set_error(SKM_ERR_INVALID_ARG, "RBQ1 needs nx2, F, popx and m");
     }
+    if ((x->flags & SKM_FLAG_SYMMETRIC) && x->repr != SKM_REPR_RBQ1)
+        return set_error(SKM_ERR_INVALID_ARG, "SKM_FLAG_SYMMETRIC applies to RBQ1 only");
     if (x->repr == SKM_REPR_LVQ4) {
         if (x->n > MAX_N_LVQ4)
             return set_error(SKM_ERR_UNSUPPORTED, "LVQ4 supports n <= 2^26 (got %lld)", (long long)x->n);
@@ -234,6 +236,11 @@ static int do_assign(const skm_data *x, const void *C, int k, const int32_t *pre
     case SKM_REPR_RBQ1:
         if (d <= TC_RBQ1_MAX_D) {
             SKM_TRY(tc_assign_rbq1(x, static_cast<const float *>(C), k, assign, dist, b.tc, st));
+        } else if (x->flags & SKM_FLAG_SYMMETRIC) {
+            uint32_t *yw = reinterpret_cast<uint32_t *>(b.planes);  // k sign words per centroid row fit
+            SKM_CUDA_TRY(launch_rbq1_cprep_sym(static_cast<const float *>(C), k, d, x->m, nullptr, 0, yw, b.info, st));
+            SKM_CUDA_TRY(launch_assign_rbq1_sym(static_cast<const uint32_t *>(x->x), x->nx2, x->F, n, d, yw, b.info, k,
+                                                assign, dist, st));
         } else {
             SKM_CUDA_TRY(launch_rbq1_cprep(static_cast<const float *>(C), k, d, x->m, b.planes,
                                            b.info, st));

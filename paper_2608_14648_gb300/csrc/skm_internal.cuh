@@ -125,6 +125,12 @@ cudaError_t launch_rbq1_cprep(const float *C, int k, int d, const float *m, uint
 inline float rbq1_isd(int d) { return (float)(1.0 / sqrt((double)d)); }
 cudaError_t launch_rbq1_cprep_tc(const float *C, int k, int d, const float *m, uint8_t *yq, int dq,
                                  Rbq1CInfo *info, cudaStream_t st);
+// symmetric 1-bit variant: binarized centroids (e4m3 +-1 codes and/or sign words)
+cudaError_t launch_rbq1_cprep_sym(const float *C, int k, int d, const float *m, uint8_t *yq, int dq, uint32_t *yw,
+                                  Rbq1CInfo *info, cudaStream_t st);
+cudaError_t launch_assign_rbq1_sym(const uint32_t *codes, const float *nx2, const float *F, int64_t n, int d,
+                                   const uint32_t *yw, const Rbq1CInfo *info, int k, int32_t *assign, float *dist,
+                                   cudaStream_t st);
 cudaError_t launch_row_sqnorm_u8(const uint8_t *codes, int64_t n, int d, int32_t *out,
                                  cudaStream_t st);
 // assignment

@@ -135,3 +135,13 @@ def test_lvq4_arguments_are_rejected_before_launch(skm):
     # hierarchical fit needs d <= 1024
     cfg = skm.HierConfig(8, 2, 1, 1, 0)
     assert L.skm_hier_workspace_size(ctypes.byref(cfg), ctypes.byref(lvq_data(d=2048))) == 0
+
+
+def test_symmetric_flag_is_validated(skm):
+    L = skm.lib()
+    x = _data(skm, repr_=1)  # SQ8
+    x.flags = skm.FLAG_SYMMETRIC
+    assert L.skm_assign(ctypes.byref(x), FAKE, 4, None, FAKE, None, FAKE, 1 << 30, None) == 1
+    r = skm.Data(skm.REPR_RBQ1, 16, 100, 0x1000, FAKE, FAKE, FAKE, FAKE, 0, skm.FLAG_SYMMETRIC)
+    assert L.skm_assign_rbq1_noalloc(ctypes.byref(r), FAKE, 4, FAKE, None, None) == 2
+    assert L.skm_workspace_size(0, ctypes.byref(r), 4) > 0

@@ -915,3 +915,32 @@ def test_assign_rbq1_extreme_code_sums_exact(skm, d):
     ao, esto = oracle.rbq1_assign(h["codes"], h["nx2"], h["F"], h["popx"], d, prep)
     np.testing.assert_array_equal(a.cpu().numpy(), ao)
     np.testing.assert_array_equal(est.cpu().numpy(), esto)
+
+
+# ------------------------------------------- symmetric 1-bit (XOR + POPCOUNT)
+@pytest.mark.parametrize("n,d,k", [(3000, 768, 300), (777, 33, 7), (1000, 1024, 65), (600, 1500, 40),
+                                   (400, 2048, 33)])
+def test_assign_rbq1_symmetric_bitexact(skm, n, d, k):
+    X = _points(n, d, seed=n + 7)
+    r = skm.skm_quantize(skm.REPR_RBQ1, X.to(DEV))
+    pts = skm.rbq1_points(r, d).with_flags(skm.FLAG_SYMMETRIC)
+    h = _rbq1_host(r)
+    C = X[synth.forgy_indices(n, k, seed=11)].clone()
+    a, est = skm.skm_assign(pts, C.to(DEV))
+    ao, eo = oracle.rbq1_assign_sym(h["codes"], h["nx2"], h["F"], d, oracle.rbq1_centroid_sym(C.numpy(), h["m"]))
+    np.testing.assert_array_equal(a.cpu().numpy(), ao)
+    np.testing.assert_array_equal(est.cpu().numpy(), eo)
+
+
+def test_fit_rbq1_symmetric_trajectory_bitexact(skm):
+    n, d, k, iters = 8000, 256, 50, 5
+    X = _points(n, d, seed=12)
+    r = skm.skm_quantize(skm.REPR_RBQ1, X.to(DEV))
+    pts = skm.rbq1_points(r, d).with_flags(skm.FLAG_SYMMETRIC)
+    idx = synth.forgy_indices(n, k, seed=12)
+    C, a, _, _, _ = skm.skm_fit(pts, k, iters, init_idx=idx.to(DEV))
+    h = _rbq1_host(r)
+    C0 = oracle.rbq1_decode_points(h["codes"], h["F"], d, h["m"], pts.rbq1_exp, idx.numpy())
+    Co, ao = oracle.lloyd_rbq1_sym(h["codes"], h["nx2"], h["F"], h["popx"], d, h["m"], C0, iters, pts.rbq1_exp)
+    np.testing.assert_array_equal(a.cpu().numpy(), ao)
+    np.testing.assert_array_equal(C.cpu().numpy(), Co)
