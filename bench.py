@@ -340,7 +340,15 @@ def run_ours(args):
         h2d = X_host.numel() * 4 + 2 * K * DIM * 4
         d2h = 2 * N_POINTS * 4 + 2 * K * DIM * 4
         e2e_steps = max(2, min(args.steps, 5))
+        # the host link's copy rate just before the run (the e2e step is bound by
+        # it; it varies with other traffic on the shared host)
         torch.cuda.synchronize()
+        p0, p1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        p0.record(stream)
+        Xd2.copy_(X_host, non_blocking=True)
+        p1.record(stream)
+        torch.cuda.synchronize()
+        h2d_probe_gbs = X_host.numel() * 4 / (p0.elapsed_time(p1) / 1e3) / 1e9
         if world > 1:
             dist.barrier()
         s0, s1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
@@ -381,6 +389,7 @@ def run_ours(args):
         e2e = {"value": world * 2.0 * N_POINTS * K * e2e_steps / (ems / 1e3), "unit": "distances/s",
                "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "steps": e2e_steps,
                "host_enqueue_ms_per_step": round(statistics.mean(host_ms), 3),
+               "h2d_probe_gbs": round(h2d_probe_gbs, 1),
                "ms_per_step": ems / e2e_steps,
                "path": f"pinned host fp32 points -> H2D in {nchunk} row ranges on a copy stream, each "
                        "range assigned (fp32) and encoded + assigned (1-bit) once it has landed -> "
