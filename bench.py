@@ -329,6 +329,7 @@ def run_ours(args):
         wsU2 = skm.workspace(skm.OP_UPDATE, probe32, K)
         copy_stream = torch.cuda.Stream()
         landed = [torch.cuda.Event() for _ in range(nchunk)]
+        c_landed = torch.cuda.Event()
         # per-range point descriptors over the fixed device buffers (views)
         pcs = [skm.Points(skm.REPR_F32, Xd2[b0:b1], DIM) for b0, b1 in bounds]
         qouts = [{"codes": codesE[b0:b1], "nx2": nx2E[b0:b1], "F": FE[b0:b1], "popx": popxE[b0:b1]}
@@ -355,13 +356,17 @@ def run_ours(args):
         s0.record(stream)
         for _ in range(e2e_steps):
             th0 = time.perf_counter()
-            copy_stream.wait_stream(stream)  # the previous step is done with Xd2
+            copy_stream.wait_stream(stream)  # the previous step is done with Xd2 and the centroids
             with torch.cuda.stream(copy_stream):
+                # centroids first: queued behind the point ranges on the same copy
+                # engine they would hold back every range's work
+                Cd32.copy_(C_host32, non_blocking=True)
+                CdR.copy_(C_hostR, non_blocking=True)
+                c_landed.record(copy_stream)
                 for (b0, b1), ev in zip(bounds, landed):
                     Xd2[b0:b1].copy_(X_host[b0:b1], non_blocking=True)
                     ev.record(copy_stream)
-            Cd32.copy_(C_host32, non_blocking=True)
-            CdR.copy_(C_hostR, non_blocking=True)
+            stream.wait_event(c_landed)
             part32e.zero_()
             cnt32e.zero_()
             for (b0, b1), ev, pc, qo, prc in zip(bounds, landed, pcs, qouts, prcs):
