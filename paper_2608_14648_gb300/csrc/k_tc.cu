@@ -66,6 +66,10 @@ constexpr int TC_CL[4] = {1, 1, 1, 1};
 // columns; 16: two buffers, the next load in flight).  Measured on GB300 at
 // 1M x 1000 x 768: 16 is 1-3% faster for both e4m3 modes.
 constexpr int F8_CW = 16;
+// The same choice for the fp32 / bf16 screen's epilogue, whose pass 1 is one
+// packed FMA per column pair: 32 is 2-4% faster there (C1 1.014 vs 1.032 ms,
+// C4 38.1 vs 39.7 ms).
+constexpr int SCR_CW = 32;
 // the e4m3 (kind::f8f6f4) modes: 128 elements per 128-byte K slice
 template <int MODE>
 constexpr bool f8_mode() { return MODE == MODE_RBQ1 || MODE == MODE_LVQ4; }
@@ -313,15 +317,6 @@ __device__ __forceinline__ float2 fmul2(float2 a, float2 b) {
         : "f"(a.x), "f"(a.y), "f"(b.x), "f"(b.y));
     return r;
 }
-__device__ __forceinline__ float2 fsub2(float2 a, float2 b) {
-    float2 r;
-    asm("{\n\t.reg .b64 ra, rb, rd;\n\t"
-        "mov.b64 ra, {%2, %3};\n\tmov.b64 rb, {%4, %5};\n\t"
-        "sub.rn.f32x2 rd, ra, rb;\n\tmov.b64 {%0, %1}, rd;\n\t}"
-        : "=f"(r.x), "=f"(r.y)
-        : "f"(a.x), "f"(a.y), "f"(b.x), "f"(b.y));
-    return r;
-}
 
 // v[i] for a lane-dependent i in [0, 32): binary select tree (no local memory).
 __device__ __forceinline__ uint32_t pick32(const uint32_t (&v)[32], int i) {
@@ -335,6 +330,24 @@ __device__ __forceinline__ uint32_t pick32(const uint32_t (&v)[32], int i) {
 #pragma unroll
     for (int t = 0; t < 2; ++t) w2[t] = (i & 2) ? w4[t + 2] : w4[t];
     return (i & 1) ? w2[1] : w2[0];
+}
+
+__device__ __forceinline__ uint32_t pick16(const uint32_t (&v)[16], int i) {
+    uint32_t w8[8], w4[4], w2[2];
+#pragma unroll
+    for (int t = 0; t < 8; ++t) w8[t] = (i & 8) ? v[t + 8] : v[t];
+#pragma unroll
+    for (int t = 0; t < 4; ++t) w4[t] = (i & 4) ? w8[t + 4] : w8[t];
+#pragma unroll
+    for (int t = 0; t < 2; ++t) w2[t] = (i & 2) ? w4[t + 2] : w4[t];
+    return (i & 1) ? w2[1] : w2[0];
+}
+template <int N>
+__device__ __forceinline__ uint32_t pickn(const uint32_t (&v)[N], int i) {
+    if constexpr (N == 32)
+        return pick32(v, i);
+    else
+        return pick16(v, i);
 }
 
 // Shared-memory matrix descriptor: K-major operand, 128-byte swizzle, rows of
@@ -638,7 +651,97 @@ __global__ void __launch_bounds__(tc_threads<NH>(), 1)
                 const uint8_t *rbuf = rec_base + b * REC_BYTES;
                 const uint32_t taddr = tmem + ((uint32_t)(q * 32) << 16) + b * BN + slice * SW;
                 const int jh = ct * BN + slice * SW;
-                if (f8_mode<MODE>()) {
+                if (MODE == MODE_SCREEN) {
+                    // chunks of SCR_CW columns (16: the next TMEM load in flight)
+                    constexpr int NC = SW / SCR_CW;
+                    constexpr int G = SCR_CW / 8;
+                    auto chunk = [&](uint32_t(&v)[SCR_CW], int c) {
+                        const int j0 = jh + c * SCR_CW;
+                        const int cc = slice * SW + c * SCR_CW;  // column offset within the tile
+                        // pass 1, two columns per packed op: s~ = ||c||^2 - 2 acc (kept in
+                        // v) and the chunk's smallest s~.  Records past k have ||c||^2 =
+                        // +inf, so s~ = +inf.
+                        float cm[G];
+#pragma unroll
+                        for (int g = 0; g < G; ++g) {
+                            cm[g] = INFINITY;
+#pragma unroll
+                            for (int i = 8 * g; i < 8 * g + 8; i += 2) {
+                                const float2 c2 = reinterpret_cast<const float2 *>(rbuf)[(cc + i) >> 1];
+                                const float2 acc = make_float2(__uint_as_float(v[i]), __uint_as_float(v[i + 1]));
+                                const float2 st = ffma2(make_float2(-2.0f, -2.0f), acc, c2);
+                                cm[g] = fminf(cm[g], fminf(st.x, st.y));
+                                v[i] = __float_as_uint(st.x);
+                                v[i + 1] = __float_as_uint(st.y);
+                            }
+                        }
+                        if (SEG && (j0 < cb || j0 + SCR_CW > ce)) {
+                            // segmented rows whose range cuts this chunk: columns
+                            // outside it do not exist for this row
+#pragma unroll
+                            for (int g = 0; g < G; ++g) {
+                                cm[g] = INFINITY;
+#pragma unroll
+                                for (int i = 8 * g; i < 8 * g + 8; ++i) {
+                                    const bool in = j0 + i >= cb && j0 + i < ce;
+                                    const float x = in ? __uint_as_float(v[i]) : INFINITY;
+                                    v[i] = __float_as_uint(x);
+                                    cm[g] = fminf(cm[g], x);
+                                }
+                            }
+                        }
+                        float cmin = cm[0];
+#pragma unroll
+                        for (int g = 1; g < G; ++g) cmin = fminf(cmin, cm[g]);
+                        sr.umin = fminf(sr.umin, cmin);
+                        const float thr = __fadd_ru(sr.umin, w2);
+                        // pass 2 (rare once the running minimum is small): pairs within
+                        // 2 W_row of the running minimum of s~ could still be the nearest
+                        if (cmin <= thr && cmin < INFINITY) {
+                            // only the 8-column groups whose minimum is inside
+                            uint32_t mask = 0;
+#pragma unroll
+                            for (int g = 0; g < G; ++g) {
+                                if (cm[g] <= thr && cm[g] < INFINITY) {
+#pragma unroll
+                                    for (int i = 8 * g; i < 8 * g + 8; ++i)
+                                        mask |= (__uint_as_float(v[i]) <= thr ? 1u : 0u) << i;
+                                }
+                            }
+                            while (mask) {
+                                const int i = __ffs(mask) - 1;
+                                mask &= mask - 1;
+                                screen_insert(sr, __uint_as_float(pickn<SCR_CW>(v, i)), j0 + i);
+                            }
+                        }
+                    };
+                    if constexpr (SCR_CW == 32) {
+#pragma unroll 1
+                        for (int c = 0; c < NC; ++c) {
+                            if (jh + c * 32 >= p.k) break;  // warp-uniform
+                            uint32_t v[32];
+                            tmem_ld32(taddr + c * 32, v);
+                            chunk(v, c);
+                        }
+                    } else if (jh < p.k) {  // warp-uniform conditions throughout
+                        uint32_t va[16], vb[16];
+                        tmem_ld16_async(taddr, va);
+                        tmem_wait16(va);
+#pragma unroll
+                        for (int c = 0; c < NC; c += 2) {
+                            const bool m1 = c + 1 < NC && jh + (c + 1) * 16 < p.k;
+                            if (m1) tmem_ld16_async(taddr + (c + 1) * 16, vb);
+                            chunk(va, c);
+                            if (!m1) break;
+                            tmem_wait16(vb);
+                            const bool m2 = c + 2 < NC && jh + (c + 2) * 16 < p.k;
+                            if (m2) tmem_ld16_async(taddr + (c + 2) * 16, va);
+                            chunk(vb, c + 1);
+                            if (!m2) break;
+                            tmem_wait16(va);
+                        }
+                    }
+                } else if (f8_mode<MODE>()) {
                     // e4m3 modes: chunks of F8_CW columns (F8_CW = 16: the next
                     // chunk's TMEM load in flight while this one is evaluated)
                     constexpr int NC = SW / F8_CW;
@@ -732,62 +835,7 @@ __global__ void __launch_bounds__(tc_threads<NH>(), 1)
                     if (j0 >= p.k) break;  // warp-uniform
                     uint32_t v[32];
                     tmem_ld32(taddr + c * 32, v);
-                    if (MODE == MODE_SCREEN) {
-                        // pass 1, two columns per packed op: s~ = ||c||^2 - 2 acc (kept in
-                        // v) and the chunk's smallest s~.  Records past k have ||c||^2 =
-                        // +inf, so s~ = +inf.
-                        float cm[4];
-#pragma unroll
-                        for (int g = 0; g < 4; ++g) {
-                            cm[g] = INFINITY;
-#pragma unroll
-                            for (int i = 8 * g; i < 8 * g + 8; i += 2) {
-                                const float2 c2 = reinterpret_cast<const float2 *>(rbuf)[(cc + i) >> 1];
-                                const float2 acc = make_float2(__uint_as_float(v[i]), __uint_as_float(v[i + 1]));
-                                const float2 st = ffma2(make_float2(-2.0f, -2.0f), acc, c2);
-                                cm[g] = fminf(cm[g], fminf(st.x, st.y));
-                                v[i] = __float_as_uint(st.x);
-                                v[i + 1] = __float_as_uint(st.y);
-                            }
-                        }
-                        if (SEG && (j0 < cb || j0 + 32 > ce)) {
-                            // segmented rows whose range cuts this chunk: columns
-                            // outside it do not exist for this row
-#pragma unroll
-                            for (int g = 0; g < 4; ++g) {
-                                cm[g] = INFINITY;
-#pragma unroll
-                                for (int i = 8 * g; i < 8 * g + 8; ++i) {
-                                    const bool in = j0 + i >= cb && j0 + i < ce;
-                                    const float x = in ? __uint_as_float(v[i]) : INFINITY;
-                                    v[i] = __float_as_uint(x);
-                                    cm[g] = fminf(cm[g], x);
-                                }
-                            }
-                        }
-                        sr.umin = fminf(sr.umin, fminf(fminf(cm[0], cm[1]), fminf(cm[2], cm[3])));
-                        const float thr = __fadd_ru(sr.umin, w2);
-                        // pass 2 (rare once the running minimum is small): pairs within
-                        // 2 W_row of the running minimum of s~ could still be the nearest
-                        const float cmin = fminf(fminf(cm[0], cm[1]), fminf(cm[2], cm[3]));
-                        if (cmin <= thr && cmin < INFINITY) {
-                            // only the 8-column groups whose minimum is inside
-                            uint32_t mask = 0;
-#pragma unroll
-                            for (int g = 0; g < 4; ++g) {
-                                if (cm[g] <= thr && cm[g] < INFINITY) {
-#pragma unroll
-                                    for (int i = 8 * g; i < 8 * g + 8; ++i)
-                                        mask |= (__uint_as_float(v[i]) <= thr ? 1u : 0u) << i;
-                                }
-                            }
-                            while (mask) {
-                                const int i = __ffs(mask) - 1;
-                                mask &= mask - 1;
-                                screen_insert(sr, __uint_as_float(pick32(v, i)), j0 + i);
-                            }
-                        }
-                    } else if (MODE == MODE_SQ8) {
+                    if (MODE == MODE_SQ8) {
 #pragma unroll
                         for (int i = 0; i < 32; ++i) {
                             const int32_t dot = __float2int_rn(__uint_as_float(v[i]));
