@@ -332,7 +332,7 @@ __device__ __forceinline__ uint32_t pick32(const uint32_t (&v)[32], int i) {
     return (i & 1) ? w2[1] : w2[0];
 }
 
-__device__ __forceinline__ uint32_t pick16(const uint32_t (&v)[16], int i) {
+__device__ __forceinline__ __attribute__((unused)) uint32_t pick16(const uint32_t (&v)[16], int i) {
     uint32_t w8[8], w4[4], w2[2];
 #pragma unroll
     for (int t = 0; t < 8; ++t) w8[t] = (i & 8) ? v[t + 8] : v[t];
