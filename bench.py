@@ -580,6 +580,42 @@ def _run_hier(args, name, n, k, idx, runs):
         torch.cuda.empty_cache()
 
 
+def _quality(args, name, X, idx, k, runs, sq8_q):
+    """Clustering quality in full precision: every representation's fit (the
+    configured iterations from the same Forgy indices) evaluated on the raw
+    fp32 points -- WCSS = sum ||x - c_a||^2 with SQ8 centroids decoded -- next
+    to the fp32 fit's."""
+    import paper_2608_14648_gb300 as skm
+
+    d = X.shape[1]
+    p32 = skm.Points(skm.REPR_F32, X, d)
+    C32, a32, _, _, _ = skm.skm_fit(p32, k, args.iters, init_idx=idx, want_objective=False, want_dist=False)
+    w32 = skm.skm_objective(X, C32, a32)
+    out = {"config": args.config, "workload": name, "quality": "full-precision WCSS after the fit",
+           "iters": args.iters, "fp32_wcss": w32}
+    for label, pts, _, _, _, _ in runs:
+        if label in ("fp32",) or label.endswith("_prune") or label.endswith("_symmetric"):
+            continue
+        C, a, _, _, _ = skm.skm_fit(pts, k, args.iters, init_idx=idx, want_objective=False, want_dist=False)
+        if label == "sq8":
+            C = skm.skm_sq8_decode(C, sq8_q["b"], sq8_q["s"])
+        w = skm.skm_objective(X, C, a)
+        out[f"{label}_wcss"] = w
+        out[f"{label}_vs_fp32"] = round(w / w32, 6)
+        if label == "rbq1" and args.iters > 0:
+            # Section 4 ("Closing RabitQ's Gap in Balance"): the last update from
+            # the raw vectors with the quantized run's assignment, then a final
+            # quantized assignment
+            C, a, _, _, _ = skm.skm_fit(pts, k, args.iters - 1, init_idx=idx, want_objective=False,
+                                        want_dist=False)
+            C, _ = skm.skm_update(p32, a, C)
+            a, _ = skm.skm_assign(pts, C, want_dist=False)
+            w = skm.skm_objective(X, C, a)
+            out["rbq1_raw_last_update_wcss"] = w
+            out["rbq1_raw_last_update_vs_fp32"] = round(w / w32, 6)
+    print(json.dumps(out), flush=True)
+
+
 def run_config(args):
     """One JSON line per representation of a workload configuration: the
     median over Lloyd iterations 2..iters of (centroid prep + assign + update)
@@ -618,9 +654,10 @@ def run_config(args):
         pL = skm.lvq4_points(skm.skm_quantize(skm.REPR_LVQ4, X), spec.d).with_screen()
         CL, _, _, _, _ = skm.skm_fit(pL, k, 0, init_idx=idx, want_objective=False, want_dist=False)
         runs.append(("lvq4", pL, CL, spec.d, 2 * bf16_peak, "e4m3"))
+    sq8_q = None
     if args.config == "c2":
         q = skm.skm_quantize(skm.REPR_SQ8, X)
-        del X
+        sq8_q = q
         runs.append(("sq8", skm.Points(skm.REPR_SQ8, q["codes"], spec.d).with_screen(),
                      q["codes"][idx].clone(), spec.d, bf16_peak, "bf16"))
         if args.prune:
@@ -652,6 +689,8 @@ def run_config(args):
     if args.hier:
         _run_hier(args, name, n, k, idx, runs)
         return
+    if args.config in ("c1", "c2"):
+        _quality(args, name, X, idx, k, runs, sq8_q)
     for label, pts, C, d, peak, kind in runs:
         C = C.clone()
         wsA = skm.workspace(skm.OP_ASSIGN, pts, k)
