@@ -580,6 +580,36 @@ def _run_hier(args, name, n, k, idx, runs):
         torch.cuda.empty_cache()
 
 
+def _timed_projection(args, name, X, P, mean, out_dtype, peaks):
+    """skm_project on the tensor cores (timed with CUDA events, after one
+    warm-up call) and once on CUDA cores for comparison; returns Y."""
+    import torch
+
+    import paper_2608_14648_gb300 as skm
+
+    n, d = X.shape
+    dout = P.shape[1]
+    Y = skm.skm_project(X, P, mean, out_dtype=out_dtype)
+    ev = [torch.cuda.Event(enable_timing=True) for _ in range(4)]
+    ev[0].record()
+    Y = skm.skm_project(X, P, mean, out_dtype=out_dtype)
+    ev[1].record()
+    torch.cuda.synchronize()
+    t_tc = ev[0].elapsed_time(ev[1])
+    ev[2].record()
+    skm.skm_project(X, P, mean, out_dtype=out_dtype, cuda_cores=True)
+    ev[3].record()
+    torch.cuda.synchronize()
+    t_cc = ev[2].elapsed_time(ev[3])
+    work = 6 * 2.0 * n * d * dout  # bf16 tensor flop: six part products
+    print(json.dumps({"config": args.config, "workload": name, "projection": f"{n} x {d} -> {dout}",
+                      "tensor_ms": round(t_tc, 3), "cuda_core_ms": round(t_cc, 3),
+                      "tensor_tflops": round(work / (t_tc / 1e3) / 1e12, 1),
+                      "frac_of_bf16_peak": round(work / (t_tc / 1e3) / 1e12 / peaks["bf16_tflops"], 4),
+                      "note": "includes the bf16 split pass (HBM) and the six-product GEMM"}), flush=True)
+    return Y
+
+
 def _quality(args, name, X, idx, k, runs, sq8_q):
     """Clustering quality in full precision: every representation's fit (the
     configured iterations from the same Forgy indices) evaluated on the raw
@@ -665,7 +695,7 @@ def run_config(args):
                          q["codes"][idx].clone(), spec.d, None, "int32 CUDA cores"))
     if args.config == "c3":
         P = synth.haar_rotation(spec.d, 99).to(torch.float32).contiguous().to(dev)
-        Y = skm.skm_project(X, P)
+        Y = _timed_projection(args, name, X, P, None, skm.DTYPE_F32, peaks)
         del X
         q = skm.skm_quantize(skm.REPR_RBQ1, Y)
         if args.lvq4:
@@ -679,7 +709,7 @@ def run_config(args):
     if args.config == "c4":
         dp = 256
         mean, P, _ = skm.skm_pca_fit(X, dp)
-        Yb = skm.skm_project(X, P, mean, out_dtype=skm.DTYPE_BF16).view(torch.int16)
+        Yb = _timed_projection(args, name, X, P, mean, skm.DTYPE_BF16, peaks).view(torch.int16)
         del X
         Cb = (Yb[idx].to(torch.int32) << 16).view(torch.float32).contiguous()
         runs.append(("bf16_screen", skm.Points(skm.REPR_BF16, Yb, dp).with_screen(), Cb, dp, bf16_peak, "bf16"))

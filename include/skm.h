@@ -131,7 +131,9 @@ uint64_t skm_kernel_launches(void);
 
 /* Bytes of scratch needed by op for these points and k centroids.
  * op: 0 = skm_assign, 1 = skm_update, 2 = skm_fit, 3 = skm_quantize,
- *     4 = skm_pca_fit, 5 = skm_assign_segmented.
+ *     4 = skm_pca_fit, 5 = skm_assign_segmented, 6 = skm_project on tensor
+ *     cores in one pass (k = d_out), 7 = the smallest workspace skm_project
+ *     takes for its tensor-core path (rows in chunks of 128).
  * Returns 0 with skm_last_error() set when the arguments are invalid. */
 size_t skm_workspace_size(int op, const skm_data *x, int k);
 
@@ -143,10 +145,16 @@ size_t skm_workspace_size(int op, const skm_data *x, int k);
  *   P      float32 [d][d_out], row-major (column j = output direction j)
  *   Y      out_dtype [n][d_out]: SKM_DTYPE_F32 (float) or SKM_DTYPE_BF16
  *          (bf16 bit patterns, rounded half to even from the fp32 result)
- * fp32 arithmetic.  d_out <= d.
- * ------------------------------------------------------------------------ */
+ * fp32 accuracy.  d_out <= d.  With a workspace of at least
+ * skm_workspace_size(6, x = {n, d}, k = d_out) bytes (or the smaller minimum
+ * it reports as skm_workspace_size(7, ...), rows then go in chunks) the
+ * product runs on the tensor cores: x - mean and P are split into three bf16
+ * parts each (x = x1 + x2 + x3 exactly, each part the round-to-nearest bf16
+ * of the remainder) and the six products with i + j <= 4 are accumulated in
+ * fp32 (the three left out are below 2^-24 relative).  ws == NULL (or
+ * smaller than the minimum): an fp32 CUDA-core tile GEMM.  Asynchronous. */
 int skm_project(const float *X, int64_t n, int d, const float *mean, const float *P,
-                int d_out, int out_dtype, void *Y, void *stream);
+                int d_out, int out_dtype, void *Y, void *ws, size_t ws_bytes, void *stream);
 
 /* Unprojection of centroids found in a projected space back to the original
  * space (Section 4, "Dimensionality Reduction and Vector Search", approach 2):

@@ -104,7 +104,7 @@ def lib():
             "skm_workspace_size": ([i32, vp, i32], sz),
             "skm_screen_bytes": ([vp], sz),
             "skm_screen_prep": ([vp, vp, sz, vp], i32),
-            "skm_project": ([vp, i64, i32, vp, vp, i32, i32, vp, vp], i32),
+            "skm_project": ([vp, i64, i32, vp, vp, i32, i32, vp, vp, sz, vp], i32),
             "skm_make_rotation": ([u64, i32, vp], i32),
             "skm_project_hadamard": ([vp, i64, i32, vp, vp, i32, i32, vp, vp], i32),
             "skm_unproject": ([vp, i64, i32, vp, vp, i32, vp, vp], i32),
@@ -207,11 +207,27 @@ def skm_workspace_size(op, pts: Points, k) -> int:
     return n
 
 
-def skm_project(X, P, mean=None, out_dtype=DTYPE_F32, stream=None):
+OP_PROJECT, OP_PROJECT_MIN = 6, 7
+
+
+def skm_project(X, P, mean=None, out_dtype=DTYPE_F32, stream=None, ws=None, max_ws_bytes=None, cuda_cores=False):
+    """Y = (X - mean) P.  Tensor cores (fp32 accuracy from bf16 parts) with a
+    workspace of up to max_ws_bytes (default: one pass over all rows);
+    cuda_cores=True selects the fp32 CUDA-core kernel (no workspace)."""
     n, d = X.shape
     d_out = P.shape[1]
     Y = torch.empty(n, d_out, device=X.device, dtype=torch.float32 if out_dtype == DTYPE_F32 else torch.bfloat16)
-    _check(lib().skm_project(_ptr(X), n, d, _ptr(mean), _ptr(P), d_out, out_dtype, _ptr(Y), _stream(stream)))
+    if cuda_cores:
+        ws = None
+    elif ws is None:
+        probe = Data(REPR_F32, d, n, 0, None, None, None, None, 0, 0)
+        full = lib().skm_workspace_size(OP_PROJECT, ctypes.byref(probe), d_out)
+        need = full if max_ws_bytes is None else max(min(full, int(max_ws_bytes)),
+                                                      lib().skm_workspace_size(OP_PROJECT_MIN, ctypes.byref(probe),
+                                                                               d_out))
+        ws = _ws(need, X.device)
+    _check(lib().skm_project(_ptr(X), n, d, _ptr(mean), _ptr(P), d_out, out_dtype, _ptr(Y), _ptr(ws),
+                             0 if ws is None else ws.numel(), _stream(stream)))
     return Y
 
 

@@ -54,14 +54,21 @@ constexpr int B_STAGE = BN * BK * 2;  // 32 KiB
 constexpr int TCAND = 4;
 constexpr unsigned long long WAIT_LIMIT_NS = 2000000000ull;  // 2 s per barrier wait
 
-enum { MODE_SCREEN = 0, MODE_SQ8 = 1, MODE_RBQ1 = 2, MODE_LVQ4 = 3 };
+enum { MODE_SCREEN = 0, MODE_SQ8 = 1, MODE_RBQ1 = 2, MODE_LVQ4 = 3, MODE_GEMM = 4 };
 // epilogue warps per TMEM lane quarter, and CTAs per cluster (centroid
 // slices multicast across the cluster), by mode.  Clusters of 2 run
 // correctly but measured slower on GB300 (the pair's pipelines wait on each
 // other's slowest epilogue: fp32 0.999 vs 0.956 ms, 1-bit 0.602 vs 0.554 ms
 // at 1M x 1000 x 768), so every mode runs one CTA per cluster.
-constexpr int TC_NH[4] = {4, 2, 4, 4};
-constexpr int TC_CL[4] = {1, 1, 1, 1};
+constexpr int TC_NH[5] = {4, 2, 4, 4, 4};
+constexpr int TC_CL[5] = {1, 1, 1, 1, 1};
+// GEMM mode (the projection Y = (X - mean) P in fp32 accuracy from bf16
+// parts x = x1 + x2 + x3, P = p1 + p2 + p3): K segments of (A part, B part),
+// the smallest products first; parts i + j > 4 (below 2^-24 relative) are left
+// out.  The A parts are stacked as rows [part][n], the B parts as [part][dout].
+constexpr int GEMM_NSEG = 6;
+__device__ constexpr int GEMM_SEG_A[GEMM_NSEG] = {2, 1, 0, 1, 0, 0};
+__device__ constexpr int GEMM_SEG_B[GEMM_NSEG] = {0, 1, 2, 0, 1, 0};
 // Columns per TMEM load in the e4m3 epilogues (32: one load and wait per 32
 // columns; 16: two buffers, the next load in flight).  Measured on GB300 at
 // 1M x 1000 x 768: 16 is 1-3% faster for both e4m3 modes.
@@ -128,6 +135,10 @@ struct TcParams {
     const int32_t *seg_group;
     const int32_t *seg_base;
     int nseg;
+    // GEMM mode: Y [n][dout] (fp32, or bf16 bits when y_bf16), row stride ydout
+    void *y;
+    int y_bf16;
+    int ydout;
 };
 
 // ------------------------------------------------------------- PTX helpers
@@ -448,6 +459,7 @@ __global__ void __launch_bounds__(tc_threads<NH>(), 1)
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     volatile int32_t *abort_flag = p.counters + 2;
+    constexpr int NSEG = MODE == MODE_GEMM ? GEMM_NSEG : 1;  // K segments per job
     constexpr int KC_ELEMS = f8_mode<MODE>() ? 128 : 64;  // elements per 128-byte row
 
     if (threadIdx.x == 0) {
@@ -495,13 +507,16 @@ __global__ void __launch_bounds__(tc_threads<NH>(), 1)
                 int ct_lo, ct_hi;
                 ct_range(p, rt, ct_lo, ct_hi);
                 for (int ct = ct_lo; ct < ct_hi; ++ct)
-                    for (int kc = 0; kc < p.nkc; ++kc, ++it) {
+                    for (int kt = 0; kt < NSEG * p.nkc; ++kt, ++it) {
+                        const int seg = kt / p.nkc, kc = kt - seg * p.nkc;
+                        const int arow = (int)(rt * BM) + (NSEG > 1 ? GEMM_SEG_A[seg] * (int)p.n : 0);
+                        const int brow = ct * BN + (NSEG > 1 ? GEMM_SEG_B[seg] * p.k : 0);
                         const uint32_t s = it % STAGES, ph = (it / STAGES) & 1u;
                         if (!mbar_wait(empty_bar(s), ph ^ 1u, abort_flag)) goto producer_done;
                         mbar_expect_tx(full_bar(s), A_STAGE + B_STAGE);
-                        tma_load_2d(sA + s * A_STAGE, &tmA, kc * KC_ELEMS, (int)(rt * BM), full_bar(s));
+                        tma_load_2d(sA + s * A_STAGE, &tmA, kc * KC_ELEMS, arow, full_bar(s));
                         if (CL == 1)
-                            tma_load_2d(sB + s * B_STAGE, &tmB, kc * KC_ELEMS, ct * BN, full_bar(s));
+                            tma_load_2d(sB + s * B_STAGE, &tmB, kc * KC_ELEMS, brow, full_bar(s));
                         else
                             tma_load_2d_mc(sB + s * B_STAGE + crank * (B_STAGE / CL), &tmB, kc * KC_ELEMS,
                                            ct * BN + (int)crank * (BN / CL), full_bar(s),
@@ -521,7 +536,7 @@ __global__ void __launch_bounds__(tc_threads<NH>(), 1)
                     if (!mbar_wait(tempty_bar(b), bph ^ 1u, abort_flag)) goto mma_done;
                     tc_fence_after();
                     const uint32_t dcol = tmem + b * BN;
-                    for (int kc = 0; kc < p.nkc; ++kc, ++it) {
+                    for (int kc = 0; kc < NSEG * p.nkc; ++kc, ++it) {
                         const uint32_t s = it % STAGES, ph = (it / STAGES) & 1u;
                         if (!mbar_wait(full_bar(s), ph, abort_flag)) goto mma_done;
                         tc_fence_after();
@@ -572,7 +587,7 @@ __global__ void __launch_bounds__(tc_threads<NH>(), 1)
             } else if (f8_mode<MODE>()) {
                 if (te < 128) pre4 = __ldg(p.rinfo + ctn * 128 + te);
                 else if (te < 256) pre4 = __ldg(p.rinfoq + ctn * 128 + (te - 128));
-            } else {
+            } else if (MODE == MODE_SQ8) {
                 if (te < 256) pre1 = __ldg(p.nc + ctn * 256 + te);
             }
         };
@@ -582,7 +597,7 @@ __global__ void __launch_bounds__(tc_threads<NH>(), 1)
                 if (te < 128) reinterpret_cast<float2 *>(rb)[te] = pre2;
             } else if (f8_mode<MODE>()) {
                 if (te < 256) reinterpret_cast<float4 *>(rb)[te] = pre4;
-            } else {
+            } else if (MODE == MODE_SQ8) {
                 if (te < 256) reinterpret_cast<int32_t *>(rb)[te] = pre1;
             }
         };
@@ -633,7 +648,7 @@ __global__ void __launch_bounds__(tc_threads<NH>(), 1)
                 rf2 = __fmul_rn(-2.0f, f.y);
                 a2 = __fmul_rn(-2.0f, f.w);
                 rnx2 = f.z;
-            } else {
+            } else if (MODE == MODE_RBQ1) {
                 rnx2 = valid ? p.nx2[row] : 0.0f;
                 rf2 = valid ? __fmul_rn(-2.0f, p.F[row]) : 0.0f;  // exact
                 rpc = valid ? (float)(2 * p.popx[row] - p.d) : 0.0f;
@@ -651,7 +666,47 @@ __global__ void __launch_bounds__(tc_threads<NH>(), 1)
                 const uint8_t *rbuf = rec_base + b * REC_BYTES;
                 const uint32_t taddr = tmem + ((uint32_t)(q * 32) << 16) + b * BN + slice * SW;
                 const int jh = ct * BN + slice * SW;
-                if (MODE == MODE_SCREEN) {
+                if (MODE == MODE_GEMM) {
+                    // write the accumulator row out: 32 columns per TMEM load
+#pragma unroll 1
+                    for (int c = 0; c < SW / 32; ++c) {
+                        const int col0 = jh + c * 32;
+                        if (col0 >= p.ydout) break;  // warp-uniform
+                        uint32_t v[32];
+                        tmem_ld32(taddr + c * 32, v);
+                        if (valid) {
+                        if (p.y_bf16) {
+                            uint16_t *yr = static_cast<uint16_t *>(p.y) + row * p.ydout;
+                            if (col0 + 32 <= p.ydout && (p.ydout % 8) == 0) {
+                                uint32_t w[16];
+#pragma unroll
+                                for (int i = 0; i < 16; ++i)
+                                    w[i] = (uint32_t)__bfloat16_as_ushort(__float2bfloat16_rn(__uint_as_float(v[2 * i]))) |
+                                           ((uint32_t)__bfloat16_as_ushort(__float2bfloat16_rn(__uint_as_float(v[2 * i + 1]))) << 16);
+                                uint4 *dst = reinterpret_cast<uint4 *>(yr + col0);
+#pragma unroll
+                                for (int q4 = 0; q4 < 4; ++q4)
+                                    dst[q4] = make_uint4(w[4 * q4], w[4 * q4 + 1], w[4 * q4 + 2], w[4 * q4 + 3]);
+                            } else {
+                                for (int i = 0; i < 32 && col0 + i < p.ydout; ++i)
+                                    yr[col0 + i] = __bfloat16_as_ushort(__float2bfloat16_rn(__uint_as_float(pick32(v, i))));
+                            }
+                        } else {
+                            float *yr = static_cast<float *>(p.y) + row * p.ydout;
+                            if (col0 + 32 <= p.ydout && (p.ydout % 4) == 0) {
+                                float4 *dst = reinterpret_cast<float4 *>(yr + col0);
+#pragma unroll
+                                for (int q4 = 0; q4 < 8; ++q4)
+                                    dst[q4] = make_float4(__uint_as_float(v[4 * q4]), __uint_as_float(v[4 * q4 + 1]),
+                                                          __uint_as_float(v[4 * q4 + 2]), __uint_as_float(v[4 * q4 + 3]));
+                            } else {
+                                for (int i = 0; i < 32 && col0 + i < p.ydout; ++i)
+                                    yr[col0 + i] = __uint_as_float(pick32(v, i));
+                            }
+                        }
+                        }
+                    }
+                } else if (MODE == MODE_SCREEN) {
                     // chunks of SCR_CW columns (16: the next TMEM load in flight)
                     constexpr int NC = SW / SCR_CW;
                     constexpr int G = SCR_CW / 8;
@@ -854,6 +909,7 @@ __global__ void __launch_bounds__(tc_threads<NH>(), 1)
             // (single buffer: a publisher rewrites its slot only at the end of
             // the next point tile, after slice 0 has passed that tile's first
             // job barrier, i.e. after it has read this one)
+            if (MODE == MODE_GEMM) continue;  // no per-row reduction across slices
             if (slice > 0) {
                 uint32_t *slot = merge + ((slice - 1) * BM + rin) * MW;
                 if (MODE == MODE_SCREEN) {
@@ -1403,7 +1459,7 @@ int launch_tc(const void *xs, int64_t n, int dp, int d, const void *cs, int k, c
     // per device: the attribute and the number of clusters that fit at once
     constexpr int MAXDEV = 64;
     static std::mutex mu;
-    static int cached_clusters[4][2][MAXDEV] = {};
+    static int cached_clusters[5][2][MAXDEV] = {};
     int dev = 0;
     SKM_CUDA_TRY(cudaGetDevice(&dev));
     int max_clusters = 0;
@@ -1434,8 +1490,10 @@ int launch_tc(const void *xs, int64_t n, int dp, int d, const void *cs, int k, c
     }
     CUtensorMap ma, mb;
     const int eb = f8_mode<MODE>() ? 1 : 2;
-    SKM_TRY(make_map(&ma, xs, n, d, dp, BM, eb));
-    SKM_TRY(make_map(&mb, cs, k, d, dp, BN / CL, eb));
+    // GEMM mode: the A and B parts are stacked (rows [part][n], [part][k])
+    const int parts = MODE == MODE_GEMM ? 3 : 1;
+    SKM_TRY(make_map(&ma, xs, parts * n, d, dp, BM, eb));
+    SKM_TRY(make_map(&mb, cs, (int64_t)parts * k, d, dp, BN / CL, eb));
     TcParams p = p0;
     p.n = n;
     p.nrt = cdiv(n, BM);
@@ -1820,6 +1878,112 @@ int tc_assign_lvq4(const skm_data *x, const float *C, int k, int32_t *assign, fl
     SKM_TRY(launch_tc<MODE_LVQ4>(v.xs, n, dp, d, b.cs, k, p, st));
     add_stats_kernel<<<1, 1, 0, st>>>(b.counters, b.stats);
     SKM_CUDA_TRY(launched());
+    return SKM_OK;
+}
+
+// ------------------------------------------------------------- projection
+namespace {
+// fp32 v -> bf16 parts v1 + v2 + v3 (each the round-to-nearest-even bf16 of
+// the remainder; the remainders are exact in fp32)
+__device__ __forceinline__ void split3(float v, uint16_t &a, uint16_t &b, uint16_t &c) {
+    const __nv_bfloat16 h1 = __float2bfloat16_rn(v);
+    const float r1 = __fsub_rn(v, __bfloat162float(h1));
+    const __nv_bfloat16 h2 = __float2bfloat16_rn(r1);
+    const float r2 = __fsub_rn(r1, __bfloat162float(h2));
+    a = __bfloat16_as_ushort(h1);
+    b = __bfloat16_as_ushort(h2);
+    c = __bfloat16_as_ushort(__float2bfloat16_rn(r2));
+}
+
+// rows [0, n) of X - mean -> A parts [3][n][dp] (8 dimensions per thread)
+__global__ void proj_split_x_kernel(const float *__restrict__ X, int64_t n, int d, const float *__restrict__ mu,
+                                    int dp, uint16_t *__restrict__ A) {
+    const int no = dp / 8;
+    const int64_t total = n * no;
+    const size_t part = (size_t)n * dp;
+    for (int64_t t = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; t < total; t += (int64_t)gridDim.x * blockDim.x) {
+        const int64_t r = t / no;
+        const int i0 = (int)(t - r * no) * 8;
+        uint32_t w[3][4];
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+            uint16_t a[2], b[2], c[2];
+#pragma unroll
+            for (int u = 0; u < 2; ++u) {
+                const int i = i0 + 2 * q + u;
+                float v = 0.0f;
+                if (i < d) v = mu ? __fsub_rn(X[r * d + i], mu[i]) : X[r * d + i];
+                split3(v, a[u], b[u], c[u]);
+            }
+            w[0][q] = (uint32_t)a[0] | ((uint32_t)a[1] << 16);
+            w[1][q] = (uint32_t)b[0] | ((uint32_t)b[1] << 16);
+            w[2][q] = (uint32_t)c[0] | ((uint32_t)c[1] << 16);
+        }
+#pragma unroll
+        for (int s3 = 0; s3 < 3; ++s3)
+            *reinterpret_cast<uint4 *>(A + s3 * part + r * dp + i0) = make_uint4(w[s3][0], w[s3][1], w[s3][2], w[s3][3]);
+    }
+}
+
+// P [d][dout] -> B parts [3][dout][dp] (transposed: K-major rows per output column)
+__global__ void proj_split_p_kernel(const float *__restrict__ P, int d, int dout, int dp, uint16_t *__restrict__ B) {
+    const int64_t total = (int64_t)dout * dp;
+    const size_t part = (size_t)dout * dp;
+    for (int64_t t = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; t < total; t += (int64_t)gridDim.x * blockDim.x) {
+        const int j = (int)(t / dp), i = (int)(t - (int64_t)j * dp);
+        uint16_t a = 0, b = 0, c = 0;
+        if (i < d) split3(P[(int64_t)i * dout + j], a, b, c);
+        B[t] = a;
+        B[part + t] = b;
+        B[2 * part + t] = c;
+    }
+}
+}  // namespace
+
+size_t tc_project_ws_min(int d, int dout) {
+    const size_t dp = (size_t)round8(d);
+    return 256 + 3 * (size_t)dout * dp * 2 + 256 + 3 * (size_t)BM * dp * 2 + 256 + 64;
+}
+
+size_t tc_project_ws_full(int64_t n, int d, int dout) {
+    const size_t dp = (size_t)round8(d);
+    return 256 + 3 * (size_t)dout * dp * 2 + 256 + 3 * (size_t)n * dp * 2 + 256 + 64;
+}
+
+int tc_project(const float *X, int64_t n, int d, const float *mean, const float *P, int dout, int out_bf16, void *Y,
+               void *ws, size_t ws_bytes, cudaStream_t st) {
+    const int dp = round8(d);
+    Carver cv(ws, ws_bytes);
+    int32_t *counters = cv.take<int32_t>(16);
+    uint16_t *B = cv.take<uint16_t>((size_t)3 * dout * dp);
+    const size_t used = cv.off + 256;
+    int64_t rows = ws_bytes > used ? (int64_t)((ws_bytes - used) / ((size_t)3 * dp * 2)) : 0;
+    if (rows >= n) rows = n;
+    else rows = (rows / BM) * BM;
+    if (rows < 1) return set_error(SKM_ERR_NO_MEMORY, "projection workspace too small");
+    uint16_t *A = cv.take<uint16_t>((size_t)3 * rows * dp);
+    if (cv.off > ws_bytes) return set_error(SKM_ERR_NO_MEMORY, "projection workspace too small");
+    {
+        int64_t blocks = ((int64_t)dout * dp + 255) / 256;
+        if (blocks > 152 * 8) blocks = 152 * 8;
+        proj_split_p_kernel<<<(unsigned)blocks, 256, 0, st>>>(P, d, dout, dp, B);
+        SKM_CUDA_TRY(launched());
+    }
+    SKM_CUDA_TRY(cudaMemsetAsync(counters, 0, sizeof(int32_t) * 16, st));
+    for (int64_t r0 = 0; r0 < n; r0 += rows) {
+        const int64_t nr = n - r0 < rows ? n - r0 : rows;
+        int64_t blocks = (nr * (dp / 8) + 255) / 256;
+        if (blocks > 152 * 16) blocks = 152 * 16;
+        proj_split_x_kernel<<<(unsigned)blocks, 256, 0, st>>>(X + r0 * d, nr, d, mean, dp, A);
+        SKM_CUDA_TRY(launched());
+        TcParams p{};
+        p.counters = counters;
+        p.y = out_bf16 ? (void *)(static_cast<uint16_t *>(Y) + r0 * dout) : (void *)(static_cast<float *>(Y) + r0 * dout);
+        p.y_bf16 = out_bf16;
+        p.ydout = dout;
+        p.d = d;
+        SKM_TRY(launch_tc<MODE_GEMM>(A, nr, dp, d, B, dout, p, st));
+    }
     return SKM_OK;
 }
 

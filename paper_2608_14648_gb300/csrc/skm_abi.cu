@@ -389,6 +389,14 @@ size_t skm_workspace_size(int op, const skm_data *x, int k) {
         cv.take<int>(1);
         break;
     }
+    case 6:  // skm_project on tensor cores, one pass
+    case 7: {  // ... the smallest workspace (rows in chunks)
+        if (!x || x->d < 1 || x->d > MAX_D || x->n < 1 || k < 1 || k > x->d) {
+            set_error(SKM_ERR_INVALID_ARG, "bad skm_data / d_out for op %d", op);
+            return 0;
+        }
+        return op == 6 ? tc_project_ws_full(x->n, x->d, k) : tc_project_ws_min(x->d, k);
+    }
     case 4: {  // pca
         if (!x || x->d < 1 || x->d > MAX_D) {
             set_error(SKM_ERR_INVALID_ARG, "bad skm_data for op 4");
@@ -409,13 +417,17 @@ size_t skm_workspace_size(int op, const skm_data *x, int k) {
 }
 
 int skm_project(const float *X, int64_t n, int d, const float *mean, const float *P, int d_out,
-                int out_dtype, void *Y, void *stream) {
+                int out_dtype, void *Y, void *ws, size_t ws_bytes, void *stream) {
     if (!X || !P || !Y) return set_error(SKM_ERR_INVALID_ARG, "NULL pointer");
     if (n < 1 || d < 1 || d > MAX_D || d_out < 1 || d_out > d)
         return set_error(SKM_ERR_INVALID_ARG, "bad shape n=%lld d=%d d_out=%d", (long long)n, d,
                          d_out);
     if (out_dtype != SKM_DTYPE_F32 && out_dtype != SKM_DTYPE_BF16)
         return set_error(SKM_ERR_INVALID_ARG, "bad out_dtype %d", out_dtype);
+    if (ws && ((uintptr_t)ws & 255) != 0)
+        return set_error(SKM_ERR_INVALID_ARG, "workspace must be 256-byte aligned");
+    if (ws && ws_bytes >= tc_project_ws_min(d, d_out) && n < (int64_t(1) << 29))
+        return tc_project(X, n, d, mean, P, d_out, out_dtype == SKM_DTYPE_BF16, Y, ws, ws_bytes, S(stream));
     SKM_CUDA_TRY(launch_project(X, n, d, mean, P, d_out, out_dtype == SKM_DTYPE_BF16, Y,
                                 S(stream)));
     return SKM_OK;

@@ -63,6 +63,13 @@ int tc_assign_rbq1(const skm_data *x, const float *C, int k, int32_t *assign, fl
 // LVQ4 on tensor cores (e4m3 codes, exact integer P, Eq. final:lvq epilogue).
 int tc_assign_lvq4(const skm_data *x, const float *C, int k, int32_t *assign, float *dist,
                    TcAssignBufs &b, cudaStream_t st, const TcSeg *seg = nullptr);
+// Y = (X - mean) P on tensor cores with fp32 accuracy (bf16 parts, six
+// products); ws: at least tc_project_ws_min (rows are then processed in chunks),
+// tc_project_ws_full for one pass.
+size_t tc_project_ws_min(int d, int dout);
+size_t tc_project_ws_full(int64_t n, int d, int dout);
+int tc_project(const float *X, int64_t n, int d, const float *mean, const float *P, int dout, int out_bf16, void *Y,
+               void *ws, size_t ws_bytes, cudaStream_t st);
 // Copies the cumulative statistics; returns SKM_ERR_TIMEOUT if a pipeline
 // wait gave up.  Synchronises the stream.
 int tc_read_stats(const TcAssignBufs &b, skm_stats *st_host, cudaStream_t st);

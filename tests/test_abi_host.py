@@ -77,9 +77,14 @@ def test_invalid_arguments_are_rejected_before_launch(skm):
     rc = L.skm_fit(ctypes.byref(cfg), ctypes.byref(x), None, None, FAKE, FAKE, None, None, None, FAKE, 1 << 30, None)
     assert rc == 1
     # projection to more dims than the input
-    assert L.skm_project(FAKE, 10, 8, None, FAKE, 9, 0, FAKE, None) == 1
+    assert L.skm_project(FAKE, 10, 8, None, FAKE, 9, 0, FAKE, None, 0, None) == 1
+    # misaligned projection workspace
+    assert L.skm_project(FAKE, 10, 8, None, FAKE, 4, 0, FAKE, ctypes.c_void_p(0x1010), 1 << 20, None) == 1
+    # projection workspace sizes: one pass >= the chunked minimum
+    x8 = _data(skm, n=100000, d=64)
+    assert L.skm_workspace_size(6, ctypes.byref(x8), 32) >= L.skm_workspace_size(7, ctypes.byref(x8), 32) > 0
     # unknown workspace op
-    assert L.skm_workspace_size(7, ctypes.byref(x), 4) == 0
+    assert L.skm_workspace_size(9, ctypes.byref(x), 4) == 0
     # unknown empty-cluster policy
     cfg = skm.FitConfig(4, 3, 7)
     rc = L.skm_fit(ctypes.byref(cfg), ctypes.byref(x), FAKE, None, FAKE, FAKE, None, None, None, FAKE, 1 << 30, None)

@@ -306,16 +306,21 @@ def test_fit_rbq1_trajectory_bitexact(skm):
 
 
 # ------------------------------------------------------ projection and bf16
-@pytest.mark.parametrize("n,d,dout", [(1000, 128, 128), (777, 100, 33), (2048, 1024, 256)])
-def test_project_vs_oracle(skm, n, d, dout):
+@pytest.mark.parametrize("n,d,dout,path", [(1000, 128, 128, "tc"), (777, 100, 33, "tc"), (2048, 1024, 256, "tc"),
+                                          (3000, 96, 96, "chunked"), (777, 100, 33, "cuda_cores"),
+                                          (1000, 768, 768, "tc"), (129, 8, 3, "tc")])
+def test_project_vs_oracle(skm, n, d, dout, path):
+    """Tensor-core projection (bf16 parts, six products, one pass or in row
+    chunks) and the CUDA-core kernel: fp32 accuracy against the fp64 oracle."""
     X = _points(n, d, seed=d)
     P = synth.haar_rotation(d, 4)[:, :dout].to(torch.float32).contiguous()
     mu = X.mean(0)
-    Y = skm.skm_project(X.to(DEV), P.to(DEV), mu.to(DEV))
+    kw = {"cuda_cores": True} if path == "cuda_cores" else ({"max_ws_bytes": 1} if path == "chunked" else {})
+    Y = skm.skm_project(X.to(DEV), P.to(DEV), mu.to(DEV), **kw)
     Yo = oracle.project(X.numpy(), P.numpy(), mu.numpy())
     scale = np.linalg.norm(X.numpy() - mu.numpy(), axis=1)[:, None]
     assert np.max(np.abs(Y.cpu().numpy() - Yo) / scale) < 2e-6
-    Yb = skm.skm_project(X.to(DEV), P.to(DEV), mu.to(DEV), out_dtype=skm.DTYPE_BF16)
+    Yb = skm.skm_project(X.to(DEV), P.to(DEV), mu.to(DEV), out_dtype=skm.DTYPE_BF16, **kw)
     yb = Yb.view(torch.int16).cpu().numpy().view(np.uint16)
     ybo = oracle.round_bf16(Yo)
     # bf16 of the fp32 result vs the fp64 result: within half a bf16 ulp of
