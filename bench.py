@@ -492,6 +492,19 @@ def run_case(args):
     torch.cuda.set_device(0)
     n, d, k = args.n, args.d, args.k
     X = synth.gmm_points(n, d, max(2 * k, 16), seed=0, device="cuda")
+    if args.case == "project":  # Y = X P on tensor cores (k = output dimensions)
+        P = synth.haar_rotation(d, 1)[:, :k].to(torch.float32).contiguous().cuda()
+        skm.skm_project(X, P)
+        torch.cuda.synchronize()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record()
+        for _ in range(args.reps):
+            skm.skm_project(X, P)
+        e1.record()
+        torch.cuda.synchronize()
+        print(json.dumps({"case": "project", "n": n, "d": d, "d_out": k, "reps": args.reps,
+                          "ms_per_call": e0.elapsed_time(e1) / args.reps}))
+        return
     C = X[synth.forgy_indices(n, k, seed=0).cuda()].clone()
     if args.case in ("assign_f32", "update_f32"):
         pts = skm.Points(skm.REPR_F32, X, d).with_screen()
@@ -774,7 +787,7 @@ def main():
     ap.add_argument("--case", default=None,
                     help="single-operation run for profiling: assign_f32|assign_rbq1|assign_sq8|assign_lvq4|"
                          "assign_rbq1_popcount|assign_prune|assign_prune_sq8|update_f32|update_rbq1|update_sq8|"
-                         "update_lvq4")
+                         "update_lvq4|project")
     ap.add_argument("--n", type=int, default=200_000)
     ap.add_argument("--d", type=int, default=768)
     ap.add_argument("--k", type=int, default=1000)
