@@ -487,9 +487,15 @@ __global__ void __launch_bounds__(RS_THREADS) ring_sum_sq8_kernel(
 
 // ------------------------------------------------------------- LVQ4 rows
 // T[c][i] += Sq code_i (the fused decode-average of Section 3.1 "LVQ4"),
-// T[c][d] += Bq.  Lane l holds nibble words l + 32 t (t < NW), i.e. 8
-// dimensions per word, each with an int64 accumulator (Sq < 2^32, code < 16:
-// one 32 x 32 -> 64-bit multiply-add per row and dimension).
+// T[c][d] += Bq.  Lane l holds nibble words l + 32 t (t < NW), 8 dimensions
+// each.  Rows are taken in pairs of the same cluster: the two weights are
+// split into 16-bit halves (lo = Sq & 0xffff, hi = Sq >> 16), the two rows'
+// nibbles of two dimensions are interleaved into one word of bytes by a byte
+// permute, and __dp2a adds lo_a x_a + lo_b x_b (and the same with hi) into
+// 32-bit sums per dimension: about 1.6 instructions per row and dimension.  A
+// row without a partner of its cluster pairs with a zero weight.  Inside a run
+// of at most RS_ROWS rows the sums stay below 128 x 65535 x 15 < 2^32; the
+// flush adds lo + hi 2^16 to the int64 accumulator.
 template <int NW>
 struct Lvq4Cons {
     const int32_t *scl;
@@ -497,7 +503,10 @@ struct Lvq4Cons {
     const int64_t *bqs;   // Bq in sorted order
     unsigned long long *T;
     int d, W;
-    unsigned long long acc[8 * NW];
+    uint32_t alo[8 * NW], ahi[8 * NW];
+    uint32_t pw[NW];  // the row waiting for a partner
+    uint32_t psq;
+    bool pend;
     int64_t usum;
     int cur;
     int64_t q0;
@@ -511,17 +520,56 @@ struct Lvq4Cons {
 #pragma unroll
             for (int j = 0; j < 8; ++j) {
                 const int col = 8 * (lane + 32 * t) + j;
-                if (col < d && acc[8 * t + j]) atomicAdd(T + (int64_t)c * (d + 1) + col, acc[8 * t + j]);
-                acc[8 * t + j] = 0ull;
+                const unsigned long long v =
+                    (unsigned long long)alo[8 * t + j] + ((unsigned long long)ahi[8 * t + j] << 16);
+                if (col < d && v) atomicAdd(T + (int64_t)c * (d + 1) + col, v);
+                alo[8 * t + j] = 0u;
+                ahi[8 * t + j] = 0u;
             }
         if (lane == 0 && usum) atomicAdd(T + (int64_t)c * (d + 1) + d, (unsigned long long)usum);
         usum = 0;
+    }
+    // rows a (words xa, weight sa) and b (xb, sb) of the current cluster
+    __device__ __forceinline__ void pair(const uint32_t (&xa)[NW], uint32_t sa, const uint32_t (&xb)[NW], uint32_t sb) {
+        const uint32_t wlo = (sa & 0xffffu) | (sb << 16);
+        const uint32_t whi = (sa >> 16) | (sb & 0xffff0000u);
+#pragma unroll
+        for (int t = 0; t < NW; ++t) {
+            const uint32_t ea = xa[t] & 0x0f0f0f0fu, oa = (xa[t] >> 4) & 0x0f0f0f0fu;
+            const uint32_t eb = xb[t] & 0x0f0f0f0fu, ob = (xb[t] >> 4) & 0x0f0f0f0fu;
+            const uint32_t m02 = __byte_perm(ea, eb, 0x5140), m46 = __byte_perm(ea, eb, 0x7362);
+            const uint32_t m13 = __byte_perm(oa, ob, 0x5140), m57 = __byte_perm(oa, ob, 0x7362);
+            uint32_t *lo = alo + 8 * t, *hi = ahi + 8 * t;
+            lo[0] = __dp2a_lo(wlo, m02, lo[0]);
+            lo[2] = __dp2a_hi(wlo, m02, lo[2]);
+            lo[4] = __dp2a_lo(wlo, m46, lo[4]);
+            lo[6] = __dp2a_hi(wlo, m46, lo[6]);
+            lo[1] = __dp2a_lo(wlo, m13, lo[1]);
+            lo[3] = __dp2a_hi(wlo, m13, lo[3]);
+            lo[5] = __dp2a_lo(wlo, m57, lo[5]);
+            lo[7] = __dp2a_hi(wlo, m57, lo[7]);
+            hi[0] = __dp2a_lo(whi, m02, hi[0]);
+            hi[2] = __dp2a_hi(whi, m02, hi[2]);
+            hi[4] = __dp2a_lo(whi, m46, hi[4]);
+            hi[6] = __dp2a_hi(whi, m46, hi[6]);
+            hi[1] = __dp2a_lo(whi, m13, hi[1]);
+            hi[3] = __dp2a_hi(whi, m13, hi[3]);
+            hi[5] = __dp2a_lo(whi, m57, hi[5]);
+            hi[7] = __dp2a_hi(whi, m57, hi[7]);
+        }
+    }
+    __device__ __forceinline__ void single() {  // the waiting row with a zero-weight partner
+        const uint32_t zero[NW] = {};
+        pair(pw, psq, zero, 0u);
+        pend = false;
     }
     __device__ __forceinline__ void start(int64_t q0_, int cnt_, int lane) {
         q0 = q0_;
         cnt = cnt_;
 #pragma unroll
-        for (int t = 0; t < 8 * NW; ++t) acc[t] = 0ull;
+        for (int t = 0; t < 8 * NW; ++t) alo[t] = ahi[t] = 0u;
+        pend = false;
+        psq = 0u;
         usum = 0;
         clw = lane < cnt ? __ldg(scl + q0 + lane) : -1;
         cln = 32 + lane < cnt ? __ldg(scl + q0 + 32 + lane) : -1;
@@ -544,23 +592,33 @@ struct Lvq4Cons {
         const int c = __shfl_sync(0xffffffffu, clw, i & 31);
         const uint32_t sq = __shfl_sync(0xffffffffu, sqw, i & 31);
         const int64_t bq = __shfl_sync(0xffffffffu, bqw, i & 31);
-        if (c != cur) {
+        if (c != cur) {  // warp-uniform
+            if (pend) single();
             flush(cur, lane);
             cur = c;
         }
         usum += bq;
         const uint32_t *words = reinterpret_cast<const uint32_t *>(slot);
+        uint32_t x[NW];
 #pragma unroll
         for (int t = 0; t < NW; ++t) {
             const int w = lane + 32 * t;
-            if (w < W) {
-                const uint32_t v = words[w];
+            x[t] = w < W ? words[w] : 0u;
+        }
+        if (pend) {
+            pair(pw, psq, x, sq);
+            pend = false;
+        } else {
 #pragma unroll
-                for (int j = 0; j < 8; ++j) acc[8 * t + j] += (unsigned long long)sq * ((v >> (4 * j)) & 15u);
-            }
+            for (int t = 0; t < NW; ++t) pw[t] = x[t];
+            psq = sq;
+            pend = true;
         }
     }
-    __device__ __forceinline__ void finish(int lane) { flush(cur, lane); }
+    __device__ __forceinline__ void finish(int lane) {
+        if (pend) single();
+        flush(cur, lane);
+    }
 };
 
 template <int NW>
