@@ -219,6 +219,29 @@ def run_ours(args):
     for _ in range(args.warmup):
         step(False)
     torch.cuda.synchronize()
+    # One GPU: the step (both Lloyd iterations, every kernel of assign and
+    # update) is captured once in a CUDA graph and replayed, so no host launch
+    # gap sits between kernels; the library's launch counter during the
+    # capture gives the kernels per step.  Several GPUs: eager (the exchange is
+    # an NCCL all-reduce between the ranks).
+    graph, launches_per_step, graph_note = None, None, None
+    if world == 1 and not args.eager:
+        try:
+            side = torch.cuda.Stream()
+            side.wait_stream(stream)
+            with torch.cuda.stream(side):
+                step(False)
+            stream.wait_stream(side)
+            torch.cuda.synchronize()
+            l0 = skm.skm_kernel_launches()
+            graph = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(graph):
+                step(False)
+            launches_per_step = skm.skm_kernel_launches() - l0
+            graph.replay()
+            torch.cuda.synchronize()
+        except Exception as exc:
+            graph, graph_note = None, f"graph capture failed, eager steps: {exc!r}"[:200]
     if world > 1:
         dist.barrier()
     clocks = ClockSampler(local_rank)
@@ -228,12 +251,20 @@ def run_ours(args):
     t_start, t_end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     t_start.record(stream)
     for _ in range(args.steps):
-        step(True)
+        if graph is not None:
+            graph.replay()
+        else:
+            step(True)
     t_end.record(stream)
     torch.cuda.synchronize()
     if world > 1:
         dist.barrier()
-    launches = skm.skm_kernel_launches() - launches0
+    launches = (launches_per_step * args.steps if graph is not None
+                else skm.skm_kernel_launches() - launches0)
+    if graph is not None:  # per-kernel event times from eager steps after the timed region
+        for _ in range(3):
+            step(True)
+        torch.cuda.synchronize()
     clk = clocks.stop()
     ms = t_start.elapsed_time(t_end)
     if world > 1:
@@ -420,6 +451,8 @@ def run_ours(args):
             "config": {"workload": WORKLOAD, "n": N_POINTS, "d": DIM, "k": K, "reprs": ["f32", "rbq1"],
                        "step": "one Lloyd iteration (assign + update) per representation",
                        "l2": "inputs larger than L2 (3.1 GB fp32 points streamed every step)",
+                       "timing": ("replays of one CUDA graph capturing the whole step" if graph is not None
+                                  else "eager steps") + (f" ({graph_note})" if graph_note else ""),
                        "parallelism": f"dp{world}"},
             "roofline": roofline, "kernels": kernels, "cpu_baseline": cpu, "e2e": e2e, "clocks": clk,
             "gpu_launches": int(launches),
@@ -759,9 +792,44 @@ def run_config(args):
         t_a = float(np.median(ta[sel]))
         t_u = float(np.median(tu[sel]))
         t_it = float(np.median([x + y for x, y in zip(ta[sel], tu[sel])]))
+        # the same iteration captured once in a CUDA graph and replayed (no
+        # host launch overhead between the kernels: what small problems need)
+        t_graph, graph_note = None, None
+        try:
+            prev_buf = a.clone() if label.endswith("_prune") else None
+            side = torch.cuda.Stream()
+            side.wait_stream(stream)
+            with torch.cuda.stream(side):
+                skm.skm_assign(pts, C, k, prev_assign=prev_buf, want_dist=False, ws=wsA, out=a)
+                skm.skm_update(pts, a, C, counts=cnt, ws=wsU)
+            stream.wait_stream(side)
+            torch.cuda.synchronize()
+            graph = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(graph):
+                skm.skm_assign(pts, C, k, prev_assign=prev_buf, want_dist=False, ws=wsA, out=a)
+                if prev_buf is not None:
+                    prev_buf.copy_(a)
+                skm.skm_update(pts, a, C, counts=cnt, ws=wsU)
+            tg = []
+            for _ in range(max(iters, 2)):
+                g0, g1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+                g0.record(stream)
+                graph.replay()
+                g1.record(stream)
+                torch.cuda.synchronize()
+                tg.append(g0.elapsed_time(g1))
+            t_graph = float(np.median(tg[1:]))
+            del graph
+        except Exception as exc:  # report instead of failing the run
+            graph_note = f"graph capture failed: {exc!r}"[:200]
         out = {"config": args.config, "workload": name, "repr": label, "n": n, "d": d, "k": k,
                "iters": iters, "ms_per_iter": round(t_it, 4), "assign_ms": round(t_a, 4),
                "update_ms": round(t_u, 4), "distances_per_s": n * k / (t_it / 1e3)}
+        if t_graph is not None:
+            out["ms_per_iter_graph"] = round(t_graph, 4)
+            out["distances_per_s_graph"] = n * k / (t_graph / 1e3)
+        if graph_note:
+            out["graph_note"] = graph_note
         if peak:
             ach = 2.0 * n * k * d / (t_a / 1e3) / 1e12
             out["assign_roofline"] = {"bound": "tensor", "achieved_tflops": round(ach, 2),
@@ -784,6 +852,7 @@ def main():
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-popcount", action="store_true")
+    ap.add_argument("--eager", action="store_true", help="time eager steps instead of CUDA-graph replays")
     ap.add_argument("--case", default=None,
                     help="single-operation run for profiling: assign_f32|assign_rbq1|assign_sq8|assign_lvq4|"
                          "assign_rbq1_popcount|assign_prune|assign_prune_sq8|update_f32|update_rbq1|update_sq8|"
