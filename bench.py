@@ -538,6 +538,28 @@ def run_case(args):
         print(json.dumps({"case": "project", "n": n, "d": d, "d_out": k, "reps": args.reps,
                           "ms_per_call": e0.elapsed_time(e1) / args.reps}))
         return
+    if args.case.startswith("quantize_"):  # skm_quantize: statistics pass + encode, and encode alone
+        repr_ = {"quantize_sq8": skm.REPR_SQ8, "quantize_rbq1": skm.REPR_RBQ1,
+                 "quantize_lvq4": skm.REPR_LVQ4}[args.case]
+        ws = skm.workspace(skm.OP_QUANTIZE, skm.Points(skm.REPR_F32, X, d), 1)
+        q = skm.skm_quantize(repr_, X, ws=ws)
+        extra = {k_: q[k_] for k_ in ("b", "s", "m") if k_ in q}
+        out_t = {k_: v for k_, v in q.items() if k_ not in ("b", "s", "m")}
+        code_bytes = sum(v.numel() * v.element_size() for v in out_t.values())
+        ms = {}
+        for fit in ((False,) if repr_ == skm.REPR_LVQ4 else (True, False)):
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            torch.cuda.synchronize()
+            e0.record()
+            for _ in range(args.reps):
+                skm.skm_quantize(repr_, X, fit=fit, out=out_t, ws=ws, **extra)
+            e1.record()
+            torch.cuda.synchronize()
+            ms["fit" if fit else "encode"] = e0.elapsed_time(e1) / args.reps
+        enc_bytes = 4 * n * d + code_bytes  # read the points once, write codes and factors
+        print(json.dumps({"case": args.case, "n": n, "d": d, "reps": args.reps, "ms_per_call": ms,
+                          "encode_bytes": enc_bytes, "encode_gbs": enc_bytes / (ms["encode"] * 1e6)}))
+        return
     C = X[synth.forgy_indices(n, k, seed=0).cuda()].clone()
     if args.case in ("assign_f32", "update_f32"):
         pts = skm.Points(skm.REPR_F32, X, d).with_screen()
@@ -856,7 +878,7 @@ def main():
     ap.add_argument("--case", default=None,
                     help="single-operation run for profiling: assign_f32|assign_rbq1|assign_sq8|assign_lvq4|"
                          "assign_rbq1_popcount|assign_prune|assign_prune_sq8|update_f32|update_rbq1|update_sq8|"
-                         "update_lvq4|project")
+                         "update_lvq4|project|quantize_sq8|quantize_rbq1|quantize_lvq4")
     ap.add_argument("--n", type=int, default=200_000)
     ap.add_argument("--d", type=int, default=768)
     ap.add_argument("--k", type=int, default=1000)

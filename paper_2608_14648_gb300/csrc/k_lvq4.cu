@@ -113,6 +113,77 @@ __global__ void lvq4_encode_kernel(const float *__restrict__ X, int64_t n, int d
     }
 }
 
+// d % 4 == 0 and d <= 1024: the row stays in registers (lane l holds the
+// float4 at dimensions 128u + 4l .. + 3, all loads issued at once), so the
+// points are read once; the two lanes of a pair assemble one nibble word
+// (8 dimensions), the even lane stores it.  Same code arithmetic as
+// lvq4_encode_warp.
+constexpr int LVQ_V4 = 8;
+
+__device__ __forceinline__ uint32_t lvq4_code(float x, float lo, float s) {
+    float q = rintf(__fdiv_rn(__fsub_rn(x, lo), s));
+    q = (q >= 0.0f) ? q : 0.0f;
+    q = fminf(q, 15.0f);
+    return (uint32_t)q;
+}
+
+__global__ void lvq4_encode_v4_kernel(const float4 *__restrict__ X, int64_t n, int d, uint32_t *__restrict__ codes,
+                                      float4 *__restrict__ fac) {
+    const int lane = threadIdx.x & 31;
+    const int64_t w0 = (blockIdx.x * (int64_t)blockDim.x + threadIdx.x) >> 5;
+    const int64_t nw = ((int64_t)gridDim.x * blockDim.x) >> 5;
+    const int W = lvq4_words(d), d4 = d >> 2;
+    for (int64_t p = w0; p < n; p += nw) {
+        const float4 *x = X + p * d4;
+        float4 v[LVQ_V4];
+        float lo = INFINITY, hi = -INFINITY;
+#pragma unroll
+        for (int u = 0; u < LVQ_V4; ++u) {
+            const int j = 32 * u + lane;
+            if (j < d4) v[u] = __ldg(x + j);
+        }
+#pragma unroll
+        for (int u = 0; u < LVQ_V4; ++u) {
+            if (32 * u + lane < d4) {
+                lo = fminf(lo, fminf(fminf(v[u].x, v[u].y), fminf(v[u].z, v[u].w)));
+                hi = fmaxf(hi, fmaxf(fmaxf(v[u].x, v[u].y), fmaxf(v[u].z, v[u].w)));
+            }
+        }
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) {
+            lo = fminf(lo, __shfl_xor_sync(FULL, lo, o));
+            hi = fmaxf(hi, __shfl_xor_sync(FULL, hi, o));
+        }
+        float s = __fdiv_rn(__fsub_rn(hi, lo), 15.0f);
+        if (!(s > 0.0f)) s = 1.0f;
+        int32_t S = 0, Q = 0;
+        uint32_t *cw = codes + p * W;
+#pragma unroll
+        for (int u = 0; u < LVQ_V4; ++u) {
+            if (32 * u < d4) {  // warp-uniform
+                const int j = 32 * u + lane;
+                uint32_t h = 0;
+                if (j < d4) {
+                    const uint32_t c0 = lvq4_code(v[u].x, lo, s), c1 = lvq4_code(v[u].y, lo, s);
+                    const uint32_t c2 = lvq4_code(v[u].z, lo, s), c3 = lvq4_code(v[u].w, lo, s);
+                    S += (int32_t)(c0 + c1 + c2 + c3);
+                    Q += (int32_t)(c0 * c0 + c1 * c1 + c2 * c2 + c3 * c3);
+                    h = (c0 | (c1 << 4) | (c2 << 8) | (c3 << 12)) << (16 * (lane & 1));
+                }
+                h |= __shfl_xor_sync(FULL, h, 1);
+                const int wi = j >> 1;
+                if ((lane & 1) == 0 && wi < W) cw[wi] = h;
+            }
+        }
+        S = __reduce_add_sync(FULL, S);
+        Q = __reduce_add_sync(FULL, Q);
+        if (lane == 0) {
+            const Lvq4Vec r{lo, s, S, Q};
+            fac[p] = make_float4(r.s, r.lo, __double2float_rn(lvq4_norm(r, d)), __double2float_rn(lvq4_sum(r, d)));
+        }
+    }
+}
+
 // M = max over points of max(s, |b|) (positive floats order like their bits),
 // then e = 31 - ceil(log2 M), 0 when M == 0.
 __global__ void lvq4_maxbits_kernel(const float4 *__restrict__ fac, int64_t n, unsigned int *__restrict__ maxbits) {
@@ -370,7 +441,11 @@ __global__ void lvq4_decode_rows_kernel(const uint32_t *__restrict__ codes, cons
 }  // namespace
 
 cudaError_t launch_lvq4_encode(const float *X, int64_t n, int d, uint32_t *codes, float4 *fac, cudaStream_t st) {
-    lvq4_encode_kernel<<<grid_warps_rows(n), 256, 0, st>>>(X, n, d, codes, fac);
+    if (d % 4 == 0 && d <= 32 * 4 * LVQ_V4 && ((uintptr_t)X & 15) == 0)
+        lvq4_encode_v4_kernel<<<grid_warps_rows(n), 256, 0, st>>>(reinterpret_cast<const float4 *>(X), n, d, codes,
+                                                                   fac);
+    else
+        lvq4_encode_kernel<<<grid_warps_rows(n), 256, 0, st>>>(X, n, d, codes, fac);
     return launched();
 }
 

@@ -28,9 +28,98 @@ __global__ void colminmax_partial_kernel(const float *__restrict__ X, int64_t n,
     }
 }
 
+// d % 4 == 0: 512-thread blocks split into P row phases of G = min(d/4, 512)
+// threads; a thread owns float4 column groups g, g + G, ... over its phase's
+// contiguous part of the block's rows (four rows of loads in flight), and the
+// phases are folded in phase order through shared memory.  With the grid of
+// two blocks per SM, the bytes in flight come from 32 resident warps per SM.
+constexpr int COL_THREADS = 512;
+constexpr int COL_ROWS = 4;
+
+struct ColPhase {
+    int G, P, ph, g0;
+    int64_t a, b;  // the phase's rows [a, b)
+};
+
+__device__ __forceinline__ ColPhase col_phase(int64_t n, int d4) {
+    ColPhase c;
+    c.G = min(d4, (int)blockDim.x);
+    c.P = blockDim.x / c.G;
+    c.ph = threadIdx.x / c.G;
+    c.g0 = threadIdx.x % c.G;
+    const int64_t rows_per = (n + gridDim.x - 1) / gridDim.x;
+    const int64_t r0 = min(n, (int64_t)blockIdx.x * rows_per), r1 = min(n, r0 + rows_per);
+    const int64_t sub = (r1 - r0 + c.P - 1) / c.P;
+    c.a = min(r1, r0 + c.ph * sub);
+    c.b = min(r1, c.a + sub);
+    return c;
+}
+
+__global__ void __launch_bounds__(COL_THREADS, 2)
+    colminmax_partial_v4_kernel(const float4 *__restrict__ X, int64_t n, int d, float *__restrict__ pmin,
+                                float *__restrict__ pmax) {
+    extern __shared__ float4 col_sh[];
+    const int d4 = d >> 2;
+    const ColPhase cp = col_phase(n, d4);
+    float4 *shlo = col_sh, *shhi = col_sh + (int64_t)cp.P * d4;
+    if (cp.ph < cp.P) {
+        for (int g = cp.g0; g < d4; g += cp.G) {
+            float4 lo = make_float4(INFINITY, INFINITY, INFINITY, INFINITY);
+            float4 hi = make_float4(-INFINITY, -INFINITY, -INFINITY, -INFINITY);
+            auto take = [&](const float4 &v) {
+                lo = make_float4(fminf(lo.x, v.x), fminf(lo.y, v.y), fminf(lo.z, v.z), fminf(lo.w, v.w));
+                hi = make_float4(fmaxf(hi.x, v.x), fmaxf(hi.y, v.y), fmaxf(hi.z, v.z), fmaxf(hi.w, v.w));
+            };
+            int64_t r = cp.a;
+            for (; r + COL_ROWS <= cp.b; r += COL_ROWS) {
+                float4 v[COL_ROWS];
+#pragma unroll
+                for (int u = 0; u < COL_ROWS; ++u) v[u] = __ldg(X + (r + u) * d4 + g);
+#pragma unroll
+                for (int u = 0; u < COL_ROWS; ++u) take(v[u]);
+            }
+            for (; r < cp.b; ++r) take(__ldg(X + r * d4 + g));
+            if (cp.P == 1) {
+                reinterpret_cast<float4 *>(pmin + (int64_t)blockIdx.x * d)[g] = lo;
+                reinterpret_cast<float4 *>(pmax + (int64_t)blockIdx.x * d)[g] = hi;
+            } else {
+                shlo[cp.ph * d4 + g] = lo;
+                shhi[cp.ph * d4 + g] = hi;
+            }
+        }
+    }
+    if (cp.P == 1) return;
+    __syncthreads();
+    for (int g = threadIdx.x; g < d4; g += blockDim.x) {
+        float4 lo = shlo[g], hi = shhi[g];
+        for (int q = 1; q < cp.P; ++q) {
+            const float4 l = shlo[q * d4 + g], h = shhi[q * d4 + g];
+            lo = make_float4(fminf(lo.x, l.x), fminf(lo.y, l.y), fminf(lo.z, l.z), fminf(lo.w, l.w));
+            hi = make_float4(fmaxf(hi.x, h.x), fmaxf(hi.y, h.y), fmaxf(hi.z, h.z), fmaxf(hi.w, h.w));
+        }
+        reinterpret_cast<float4 *>(pmin + (int64_t)blockIdx.x * d)[g] = lo;
+        reinterpret_cast<float4 *>(pmax + (int64_t)blockIdx.x * d)[g] = hi;
+    }
+}
+
+// shared memory of the two phase-split column kernels: P * d4 <= 512 when
+// P > 1, so P * d <= 2048 values
+static size_t col_smem(int d, size_t per_col) {
+    const int d4 = d / 4;
+    const int G = d4 < COL_THREADS ? d4 : COL_THREADS;
+    const int P = COL_THREADS / G;
+    return P > 1 ? (size_t)P * d * per_col : 0;
+}
+
 cudaError_t launch_colminmax_partial(const float *X, int64_t n, int d, float *pmin, float *pmax,
                                      int nblk, cudaStream_t st) {
-    colminmax_partial_kernel<<<nblk, 256, 0, st>>>(X, n, d, pmin, pmax);
+    if (d % 4 == 0 && (((uintptr_t)X | (uintptr_t)pmin | (uintptr_t)pmax) & 15) == 0) {
+        const size_t sh = 2 * col_smem(d, sizeof(float));  // at most 16 KB
+        colminmax_partial_v4_kernel<<<nblk, COL_THREADS, sh, st>>>(reinterpret_cast<const float4 *>(X), n, d,
+                                                                   pmin, pmax);
+    } else {
+        colminmax_partial_kernel<<<nblk, 256, 0, st>>>(X, n, d, pmin, pmax);
+    }
     return launched();
 }
 
@@ -65,25 +154,39 @@ __device__ __forceinline__ uint32_t sq8_code(float x, float b, float s, float to
     return (uint32_t)q;
 }
 
-__global__ void sq8_encode_vec_kernel(const float4 *__restrict__ X, int64_t n16, int d,
-                                      const float *__restrict__ b, const float *__restrict__ s,
-                                      float top, uint4 *__restrict__ out) {
-    // requires d % 16 == 0: a 16-element chunk never crosses a row
-    for (int64_t t = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; t < n16;
-         t += (int64_t)gridDim.x * blockDim.x) {
-        const int c0 = (int)((t * 16) % d);
-        float4 v[4];
+// d % 4 == 0: one warp per row, lane l takes the float4 at dimensions
+// 128t + 4l .. + 3 and writes their four codes as one 32-bit word, so the
+// (b, s) loads and the code stores are contiguous across the warp; a row's
+// loads (up to SQ_V4 float4 per lane) are issued before use.
+constexpr int SQ_V4 = 8;
+
+__global__ void sq8_encode_rows_kernel(const float4 *__restrict__ X, int64_t n, int d,
+                                       const float4 *__restrict__ b, const float4 *__restrict__ s,
+                                       float top, uint32_t *__restrict__ out) {
+    const int lane = threadIdx.x & 31;
+    const int64_t warp = (blockIdx.x * (int64_t)blockDim.x + threadIdx.x) >> 5;
+    const int64_t nwarps = ((int64_t)gridDim.x * blockDim.x) >> 5;
+    const int d4 = d >> 2;
+    for (int64_t p = warp; p < n; p += nwarps) {
+        const float4 *x = X + p * d4;
+        uint32_t *o = out + p * d4;
+        for (int t0 = 0; 32 * t0 < d4; t0 += SQ_V4) {
+            float4 v[SQ_V4];
 #pragma unroll
-        for (int q = 0; q < 4; ++q) v[q] = X[t * 4 + q];
-        uint32_t w[4];
+            for (int u = 0; u < SQ_V4; ++u) {
+                const int j = 32 * (t0 + u) + lane;
+                if (j < d4) v[u] = __ldg(x + j);
+            }
 #pragma unroll
-        for (int q = 0; q < 4; ++q) {
-            const int c = c0 + 4 * q;
-            w[q] = sq8_code(v[q].x, b[c], s[c], top) | (sq8_code(v[q].y, b[c + 1], s[c + 1], top) << 8) |
-                   (sq8_code(v[q].z, b[c + 2], s[c + 2], top) << 16) |
-                   (sq8_code(v[q].w, b[c + 3], s[c + 3], top) << 24);
+            for (int u = 0; u < SQ_V4; ++u) {
+                const int j = 32 * (t0 + u) + lane;
+                if (j < d4) {
+                    const float4 bb = __ldg(b + j), ss = __ldg(s + j);
+                    o[j] = sq8_code(v[u].x, bb.x, ss.x, top) | (sq8_code(v[u].y, bb.y, ss.y, top) << 8) |
+                           (sq8_code(v[u].z, bb.z, ss.z, top) << 16) | (sq8_code(v[u].w, bb.w, ss.w, top) << 24);
+                }
+            }
         }
-        out[t] = make_uint4(w[0], w[1], w[2], w[3]);
     }
 }
 
@@ -109,10 +212,10 @@ cudaError_t launch_sq8_encode(const float *X, int64_t n, int d, const float *b, 
                               int levels, uint8_t *codes, cudaStream_t st) {
     const int64_t total = n * d;
     const float top = (float)levels;
-    if (d % 16 == 0 && (((uintptr_t)X | (uintptr_t)codes) & 15) == 0) {
-        const int64_t n16 = total / 16;
-        sq8_encode_vec_kernel<<<grid_for(n16, 256), 256, 0, st>>>(
-            reinterpret_cast<const float4 *>(X), n16, d, b, s, top, reinterpret_cast<uint4 *>(codes));
+    if (d % 4 == 0 && (((uintptr_t)X | (uintptr_t)b | (uintptr_t)s) & 15) == 0 && ((uintptr_t)codes & 3) == 0) {
+        sq8_encode_rows_kernel<<<grid_for(n * 32, 256), 256, 0, st>>>(
+            reinterpret_cast<const float4 *>(X), n, d, reinterpret_cast<const float4 *>(b),
+            reinterpret_cast<const float4 *>(s), top, reinterpret_cast<uint32_t *>(codes));
     } else {
         sq8_encode_scalar_kernel<<<grid_for(total, 256), 256, 0, st>>>(X, total, d, b, s, top, codes);
     }
@@ -169,9 +272,63 @@ __global__ void colsum_partial_kernel(const float *__restrict__ X, int64_t n, in
     }
 }
 
+// d % 4 == 0: the phase split of colminmax_partial_v4_kernel; each phase keeps
+// the Kahan recurrence per column in row order over its rows, and the phases'
+// compensated sums are added in fp64 in phase order.
+__device__ __forceinline__ void kahan_col(float &s, float &comp, float v) {
+    const float y = __fsub_rn(v, comp);
+    const float t = __fadd_rn(s, y);
+    comp = __fsub_rn(__fsub_rn(t, s), y);
+    s = t;
+}
+
+__global__ void __launch_bounds__(COL_THREADS, 2)
+    colsum_partial_v4_kernel(const float4 *__restrict__ X, int64_t n, int d, double *__restrict__ psum) {
+    extern __shared__ double col_shd[];
+    const int d4 = d >> 2;
+    const ColPhase cp = col_phase(n, d4);
+    if (cp.ph < cp.P) {
+        for (int g = cp.g0; g < d4; g += cp.G) {
+            float4 s = make_float4(0.0f, 0.0f, 0.0f, 0.0f), c = s;
+            auto take = [&](const float4 &v) {
+                kahan_col(s.x, c.x, v.x);
+                kahan_col(s.y, c.y, v.y);
+                kahan_col(s.z, c.z, v.z);
+                kahan_col(s.w, c.w, v.w);
+            };
+            int64_t r = cp.a;
+            for (; r + COL_ROWS <= cp.b; r += COL_ROWS) {
+                float4 v[COL_ROWS];
+#pragma unroll
+                for (int u = 0; u < COL_ROWS; ++u) v[u] = __ldg(X + (r + u) * d4 + g);
+#pragma unroll
+                for (int u = 0; u < COL_ROWS; ++u) take(v[u]);
+            }
+            for (; r < cp.b; ++r) take(__ldg(X + r * d4 + g));
+            double *o = cp.P == 1 ? psum + (int64_t)blockIdx.x * d + 4 * g : col_shd + (int64_t)cp.ph * d + 4 * g;
+            o[0] = (double)s.x - (double)c.x;
+            o[1] = (double)s.y - (double)c.y;
+            o[2] = (double)s.z - (double)c.z;
+            o[3] = (double)s.w - (double)c.w;
+        }
+    }
+    if (cp.P == 1) return;
+    __syncthreads();
+    for (int c = threadIdx.x; c < d; c += blockDim.x) {
+        double acc = col_shd[c];
+        for (int q = 1; q < cp.P; ++q) acc = __dadd_rn(acc, col_shd[(int64_t)q * d + c]);
+        psum[(int64_t)blockIdx.x * d + c] = acc;
+    }
+}
+
 cudaError_t launch_colsum_partial(const float *X, int64_t n, int d, double *psum, int nblk,
                                   cudaStream_t st) {
-    colsum_partial_kernel<<<nblk, 256, 0, st>>>(X, n, d, psum);
+    if (d % 4 == 0 && ((uintptr_t)X & 15) == 0) {
+        const size_t sh = col_smem(d, sizeof(double));  // at most 16 KB
+        colsum_partial_v4_kernel<<<nblk, COL_THREADS, sh, st>>>(reinterpret_cast<const float4 *>(X), n, d, psum);
+    } else {
+        colsum_partial_kernel<<<nblk, 256, 0, st>>>(X, n, d, psum);
+    }
     return launched();
 }
 
@@ -193,11 +350,14 @@ cudaError_t launch_colmean_finish(const double *psum, int nblk, int d, int64_t n
 }
 
 // ---------------------------------------------------------------------------
-// RabitQ 1-bit encode: one warp per point.  Lane l handles dimensions
-// 32w + l; the sign bits of a 32-dimension group are one __ballot_sync.
-// ||r||^2 and ||r||_1: Kahan-compensated fp32 lane sums (relative error about
-// 2^-23), then an fp64 xor-tree across lanes; F = sqrt(d) ||r||^2 / ||r||_1
-// is evaluated in fp64 and rounded once.
+// RabitQ 1-bit encode: one warp per point, r = x - m.  ||r||^2 and ||r||_1 are
+// Kahan-compensated fp32 lane sums (relative error about 2^-23); the 32 lane
+// pairs (s, -c) are folded across the warp as double-float numbers (error-free
+// TwoSum of the leading parts, trailing parts added), so the row total keeps
+// about 40 bits before its single rounding to fp32.  F = sqrt(d) ||r||^2 /
+// ||r||_1 then takes three fp32 roundings (relative error below 2^-22).  No
+// fp64 instruction runs per point: GB300 issues fp64 at a small fraction of the
+// fp32 rate, and a per-row fp64 tail bounded the former version.
 // ---------------------------------------------------------------------------
 __device__ __forceinline__ void kahan_add(float &s, float &c, float v) {
     const float y = __fsub_rn(v, c);
@@ -206,8 +366,41 @@ __device__ __forceinline__ void kahan_add(float &s, float &c, float v) {
     s = t;
 }
 
+// (hi, lo) += (h2, l2) for double-float numbers: TwoSum of the leading parts,
+// trailing parts added to the error, renormalised by FastTwoSum.
+__device__ __forceinline__ void df_add(float &hi, float &lo, float h2, float l2) {
+    const float s = __fadd_rn(hi, h2);
+    const float bb = __fsub_rn(s, hi);
+    const float e = __fadd_rn(__fsub_rn(hi, __fsub_rn(s, bb)), __fsub_rn(h2, bb));
+    const float t = __fadd_rn(e, __fadd_rn(lo, l2));
+    hi = __fadd_rn(s, t);
+    lo = __fsub_rn(t, __fsub_rn(hi, s));
+}
+
+// Folds the lane sums of one point and writes ||r||^2, F and popcount(code).
+__device__ __forceinline__ void rbq1_row_finish(float s2, float c2, float s1, float c1, int pc, int lane,
+                                                float sqrt_d, float *nx2, float *F, int32_t *popx) {
+    float h2 = s2, l2 = -c2, h1 = s1, l1 = -c1;
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+        const float a = __shfl_xor_sync(0xffffffffu, h2, o), b = __shfl_xor_sync(0xffffffffu, l2, o);
+        const float e = __shfl_xor_sync(0xffffffffu, h1, o), f = __shfl_xor_sync(0xffffffffu, l1, o);
+        df_add(h2, l2, a, b);
+        df_add(h1, l1, e, f);
+    }
+    pc = __reduce_add_sync(0xffffffffu, pc);
+    if (lane == 0) {
+        const float t2 = __fadd_rn(h2, l2), t1 = __fadd_rn(h1, l1);
+        *nx2 = t2;
+        *F = t1 > 0.0f ? __fdiv_rn(__fmul_rn(sqrt_d, t2), t1) : 0.0f;
+        *popx = pc;
+    }
+}
+
 constexpr int ENC_UNROLL = 8;
 
+// Any d: lane l takes dimensions 32w + l, the sign bits of a 32-dimension
+// group are one __ballot_sync.
 __global__ void rbq1_encode_kernel(const float *__restrict__ X, int64_t n, int d,
                                    const float *__restrict__ m, uint32_t *__restrict__ codes,
                                    float *__restrict__ nx2, float *__restrict__ F,
@@ -216,7 +409,7 @@ __global__ void rbq1_encode_kernel(const float *__restrict__ X, int64_t n, int d
     const int64_t warp = (blockIdx.x * (int64_t)blockDim.x + threadIdx.x) >> 5;
     const int64_t nwarps = ((int64_t)gridDim.x * blockDim.x) >> 5;
     const int W = (d + 31) >> 5;
-    const double sqrt_d = sqrt((double)d);
+    const float sqrt_d = __fsqrt_rn((float)d);
     for (int64_t p = warp; p < n; p += nwarps) {
         const float *x = X + p * d;
         float s2 = 0.0f, c2 = 0.0f, s1 = 0.0f, c1 = 0.0f;
@@ -244,25 +437,84 @@ __global__ void rbq1_encode_kernel(const float *__restrict__ X, int64_t n, int d
                 }
             }
         }
-        double t2 = (double)s2 - (double)c2, t1 = (double)s1 - (double)c1;
+        rbq1_row_finish(s2, c2, s1, c1, pc, lane, sqrt_d, nx2 + p, F + p, popx + p);
+    }
+}
+
+// d % 4 == 0: lane l takes the float4 at dimensions 128t + 4l .. 128t + 4l + 3,
+// so its four sign bits are bits 4(l mod 8) .. 4(l mod 8) + 3 of code word
+// 4t + l/8; an OR butterfly over each group of 8 lanes assembles the words.
+// All of a row's loads (up to ENC_V4 float4 per lane) are issued before use.
+constexpr int ENC_V4 = 8;
+
+__global__ void rbq1_encode_v4_kernel(const float4 *__restrict__ X, int64_t n, int d,
+                                      const float4 *__restrict__ m, uint32_t *__restrict__ codes,
+                                      float *__restrict__ nx2, float *__restrict__ F,
+                                      int32_t *__restrict__ popx) {
+    const int lane = threadIdx.x & 31;
+    const int64_t warp = (blockIdx.x * (int64_t)blockDim.x + threadIdx.x) >> 5;
+    const int64_t nwarps = ((int64_t)gridDim.x * blockDim.x) >> 5;
+    const int W = (d + 31) >> 5, d4 = d >> 2;
+    const float sqrt_d = __fsqrt_rn((float)d);
+    for (int64_t p = warp; p < n; p += nwarps) {
+        const float4 *x = X + p * d4;
+        float s2 = 0.0f, c2 = 0.0f, s1 = 0.0f, c1 = 0.0f;
+        int pc = 0;
+        for (int t0 = 0; 32 * t0 < d4; t0 += ENC_V4) {
+            float4 v[ENC_V4];
 #pragma unroll
-        for (int o = 16; o > 0; o >>= 1) {
-            t2 += __shfl_xor_sync(0xffffffffu, t2, o);
-            t1 += __shfl_xor_sync(0xffffffffu, t1, o);
+            for (int u = 0; u < ENC_V4; ++u) {
+                const int j = 32 * (t0 + u) + lane;
+                v[u] = j < d4 ? __ldg(x + j) : make_float4(0.0f, 0.0f, 0.0f, 0.0f);
+            }
+#pragma unroll
+            for (int u = 0; u < ENC_V4; ++u) {
+                const int t = t0 + u;
+                if (32 * t < d4) {  // warp-uniform
+                    const int j = 32 * t + lane;
+                    float4 r = make_float4(0.0f, 0.0f, 0.0f, 0.0f);
+                    if (j < d4) {
+                        const float4 mm = __ldg(m + j);
+                        r = make_float4(__fsub_rn(v[u].x, mm.x), __fsub_rn(v[u].y, mm.y),
+                                        __fsub_rn(v[u].z, mm.z), __fsub_rn(v[u].w, mm.w));
+                    }
+                    kahan_add(s2, c2, __fmul_rn(r.x, r.x));
+                    kahan_add(s2, c2, __fmul_rn(r.y, r.y));
+                    kahan_add(s2, c2, __fmul_rn(r.z, r.z));
+                    kahan_add(s2, c2, __fmul_rn(r.w, r.w));
+                    kahan_add(s1, c1, fabsf(r.x));
+                    kahan_add(s1, c1, fabsf(r.y));
+                    kahan_add(s1, c1, fabsf(r.z));
+                    kahan_add(s1, c1, fabsf(r.w));
+                    uint32_t nib = (r.x > 0.0f ? 1u : 0u) | (r.y > 0.0f ? 2u : 0u) | (r.z > 0.0f ? 4u : 0u) |
+                                   (r.w > 0.0f ? 8u : 0u);
+                    nib <<= 4 * (lane & 7);
+                    nib |= __shfl_xor_sync(0xffffffffu, nib, 1);
+                    nib |= __shfl_xor_sync(0xffffffffu, nib, 2);
+                    nib |= __shfl_xor_sync(0xffffffffu, nib, 4);
+                    const int wi = 4 * t + (lane >> 3);
+                    if ((lane & 7) == 0 && wi < W) {
+                        codes[p * W + wi] = nib;
+                        pc += __popc(nib);
+                    }
+                }
+            }
         }
-        if (lane == 0) {
-            nx2[p] = __double2float_rn(t2);
-            F[p] = (t1 > 0.0) ? __double2float_rn(__ddiv_rn(__dmul_rn(sqrt_d, t2), t1)) : 0.0f;
-            popx[p] = pc;
-        }
+        rbq1_row_finish(s2, c2, s1, c1, pc, lane, sqrt_d, nx2 + p, F + p, popx + p);
     }
 }
 
 cudaError_t launch_rbq1_encode(const float *X, int64_t n, int d, const float *m, uint32_t *codes,
                                float *nx2, float *F, int32_t *popx, cudaStream_t st) {
     const int threads = 256;
-    rbq1_encode_kernel<<<grid_for(n * 32, threads), threads, 0, st>>>(X, n, d, m, codes, nx2, F,
-                                                                      popx);
+    if (d % 4 == 0 && ((uintptr_t)X & 15) == 0 && ((uintptr_t)m & 15) == 0) {
+        rbq1_encode_v4_kernel<<<grid_for(n * 32, threads), threads, 0, st>>>(
+            reinterpret_cast<const float4 *>(X), n, d, reinterpret_cast<const float4 *>(m), codes, nx2, F,
+            popx);
+    } else {
+        rbq1_encode_kernel<<<grid_for(n * 32, threads), threads, 0, st>>>(X, n, d, m, codes, nx2, F,
+                                                                          popx);
+    }
     return launched();
 }
 

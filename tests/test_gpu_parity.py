@@ -203,7 +203,7 @@ def test_fit_f32_tiny_workload(skm):
 
 
 # ------------------------------------------------------------------ SQ8 path
-@pytest.mark.parametrize("n,d", [(2000, 64), (777, 33), (1500, 1024), (50, 1)])
+@pytest.mark.parametrize("n,d", [(2000, 64), (777, 33), (1500, 1024), (50, 1), (333, 36), (257, 1500), (5000, 772)])
 def test_quantize_sq8_bitexact(skm, n, d):
     X = _points(n, d, seed=n)
     q = skm.skm_quantize(skm.REPR_SQ8, X.to(DEV))
@@ -253,7 +253,7 @@ def _rbq1_host(r):
     return h
 
 
-@pytest.mark.parametrize("n,d", [(3000, 768), (777, 33), (500, 32), (400, 31), (100, 1)])
+@pytest.mark.parametrize("n,d", [(3000, 768), (777, 33), (500, 32), (400, 31), (100, 1), (333, 36), (257, 1500)])
 def test_encode_rbq1_vs_oracle(skm, n, d):
     X = _points(n, d, seed=n + 1)
     r = skm.skm_quantize(skm.REPR_RBQ1, X.to(DEV))
@@ -734,7 +734,8 @@ def _lvq4_host(q, d):
     return {"words": words, "codes": oracle.lvq4_unpack(words, d), "fac": q["lvq"].cpu().numpy()}
 
 
-@pytest.mark.parametrize("n,d", [(3000, 768), (777, 33), (500, 32), (400, 31), (100, 1), (300, 2048)])
+@pytest.mark.parametrize("n,d", [(3000, 768), (777, 33), (500, 32), (400, 31), (100, 1), (300, 2048), (333, 36),
+                                 (257, 1020), (100, 1024)])
 def test_encode_lvq4_bitexact(skm, n, d):
     X = _points(n, d, seed=n + 3)
     q = skm.skm_quantize(skm.REPR_LVQ4, X.to(DEV))
