@@ -95,12 +95,36 @@ __device__ __forceinline__ uint32_t pack_nibbles(uint32_t c, int lane) {
     return v;
 }
 
+// N and A (R25) take fp64 arithmetic, which GB300 issues at a small fraction
+// of its fp32 rate, and a warp instruction costs the same with one lane active
+// as with 32: a warp therefore parks the (s, b, S, Q) of 32 consecutive rows of
+// its loop in lanes 0..31 and evaluates the 32 fp64 tails together.
+struct FacBatch {
+    Lvq4Vec r{0.0f, 0.0f, 0, 0};
+    int64_t row = -1;
+    int cnt = 0;
+    __device__ __forceinline__ void put(const Lvq4Vec &v, int64_t p, int lane, float4 *fac, int d) {
+        if (lane == cnt) {
+            r = v;
+            row = p;
+        }
+        if (++cnt == 32) flush(fac, d);
+    }
+    __device__ __forceinline__ void flush(float4 *fac, int d) {
+        if (row >= 0)
+            fac[row] = make_float4(r.s, r.lo, __double2float_rn(lvq4_norm(r, d)), __double2float_rn(lvq4_sum(r, d)));
+        row = -1;
+        cnt = 0;
+    }
+};
+
 __global__ void lvq4_encode_kernel(const float *__restrict__ X, int64_t n, int d, uint32_t *__restrict__ codes,
                                    float4 *__restrict__ fac) {
     const int lane = threadIdx.x & 31;
     const int64_t w0 = (blockIdx.x * (int64_t)blockDim.x + threadIdx.x) >> 5;
     const int64_t nw = ((int64_t)gridDim.x * blockDim.x) >> 5;
     const int W = lvq4_words(d);
+    FacBatch fb;
     for (int64_t p = w0; p < n; p += nw) {
         uint32_t *cw = codes + p * W;
         const Lvq4Vec r = lvq4_encode_warp(X + p * d, d, lane, [&](int base, int ln, uint32_t c) {
@@ -108,9 +132,9 @@ __global__ void lvq4_encode_kernel(const float *__restrict__ X, int64_t n, int d
             const int wi = (base >> 3) + (ln >> 3);
             if ((ln & 7) == 0 && wi < W) cw[wi] = v;
         });
-        if (lane == 0)
-            fac[p] = make_float4(r.s, r.lo, __double2float_rn(lvq4_norm(r, d)), __double2float_rn(lvq4_sum(r, d)));
+        fb.put(r, p, lane, fac, d);
     }
+    fb.flush(fac, d);
 }
 
 // d % 4 == 0 and d <= 1024: the row stays in registers (lane l holds the
@@ -120,19 +144,31 @@ __global__ void lvq4_encode_kernel(const float *__restrict__ X, int64_t n, int d
 // lvq4_encode_warp.
 constexpr int LVQ_V4 = 8;
 
-__device__ __forceinline__ uint32_t lvq4_code(float x, float lo, float s) {
-    float q = rintf(__fdiv_rn(__fsub_rn(x, lo), s));
-    q = (q >= 0.0f) ? q : 0.0f;
-    q = fminf(q, 15.0f);
-    return (uint32_t)q;
+// clip(rint(fl((x - lo) / s)), 0, 15) with one multiplication in place of the
+// division: with rs = fl(1/s), q' = fl(a rs) (a = fl(x - lo)) is within
+// (2^-23 + 2^-24 + 2^-48) |a/s| of the correctly rounded quotient q, i.e. within
+// 2^-18.5 since a/s <= 15 / (1 - 2^-24) here (a <= fl(hi - lo), s rounded from
+// fl(hi - lo) / 15).  When q' is more than
+// 2^-17 away from every half-integer, q and q' round to the same integer;
+// otherwise (and for inf / NaN) the quotient is taken by the IEEE division.
+// The bound needs a normal rs: callers pass NaN instead of a subnormal one.
+__device__ __forceinline__ uint32_t lvq4_code(float x, float lo, float s, float rs) {
+    const float a = __fsub_rn(x, lo);
+    float q = __fmul_rn(a, rs);
+    float t = rintf(q);
+    if (!(fabsf(__fsub_rn(q, t)) < 0.5f - 0x1p-17f)) t = rintf(__fdiv_rn(a, s));
+    t = (t >= 0.0f) ? t : 0.0f;
+    t = fminf(t, 15.0f);
+    return (uint32_t)t;
 }
 
-__global__ void lvq4_encode_v4_kernel(const float4 *__restrict__ X, int64_t n, int d, uint32_t *__restrict__ codes,
+__global__ void __launch_bounds__(256, 3) lvq4_encode_v4_kernel(const float4 *__restrict__ X, int64_t n, int d, uint32_t *__restrict__ codes,
                                       float4 *__restrict__ fac) {
     const int lane = threadIdx.x & 31;
     const int64_t w0 = (blockIdx.x * (int64_t)blockDim.x + threadIdx.x) >> 5;
     const int64_t nw = ((int64_t)gridDim.x * blockDim.x) >> 5;
     const int W = lvq4_words(d), d4 = d >> 2;
+    FacBatch fb;
     for (int64_t p = w0; p < n; p += nw) {
         const float4 *x = X + p * d4;
         float4 v[LVQ_V4];
@@ -156,6 +192,8 @@ __global__ void lvq4_encode_v4_kernel(const float4 *__restrict__ X, int64_t n, i
         }
         float s = __fdiv_rn(__fsub_rn(hi, lo), 15.0f);
         if (!(s > 0.0f)) s = 1.0f;
+        float rs = __frcp_rn(s);
+        if (!(fabsf(rs) >= 0x1p-126f)) rs = __int_as_float(0x7fffffff);  // subnormal: divide every code
         int32_t S = 0, Q = 0;
         uint32_t *cw = codes + p * W;
 #pragma unroll
@@ -164,8 +202,8 @@ __global__ void lvq4_encode_v4_kernel(const float4 *__restrict__ X, int64_t n, i
                 const int j = 32 * u + lane;
                 uint32_t h = 0;
                 if (j < d4) {
-                    const uint32_t c0 = lvq4_code(v[u].x, lo, s), c1 = lvq4_code(v[u].y, lo, s);
-                    const uint32_t c2 = lvq4_code(v[u].z, lo, s), c3 = lvq4_code(v[u].w, lo, s);
+                    const uint32_t c0 = lvq4_code(v[u].x, lo, s, rs), c1 = lvq4_code(v[u].y, lo, s, rs);
+                    const uint32_t c2 = lvq4_code(v[u].z, lo, s, rs), c3 = lvq4_code(v[u].w, lo, s, rs);
                     S += (int32_t)(c0 + c1 + c2 + c3);
                     Q += (int32_t)(c0 * c0 + c1 * c1 + c2 * c2 + c3 * c3);
                     h = (c0 | (c1 << 4) | (c2 << 8) | (c3 << 12)) << (16 * (lane & 1));
@@ -177,11 +215,9 @@ __global__ void lvq4_encode_v4_kernel(const float4 *__restrict__ X, int64_t n, i
         }
         S = __reduce_add_sync(FULL, S);
         Q = __reduce_add_sync(FULL, Q);
-        if (lane == 0) {
-            const Lvq4Vec r{lo, s, S, Q};
-            fac[p] = make_float4(r.s, r.lo, __double2float_rn(lvq4_norm(r, d)), __double2float_rn(lvq4_sum(r, d)));
-        }
+        fb.put(Lvq4Vec{lo, s, S, Q}, p, lane, fac, d);
     }
+    fb.flush(fac, d);
 }
 
 // M = max over points of max(s, |b|) (positive floats order like their bits),

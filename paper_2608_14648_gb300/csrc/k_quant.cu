@@ -146,7 +146,7 @@ cudaError_t launch_sq8_params(const float *pmin, const float *pmax, int nblk, in
 }
 
 // code = clip(rint((x - b) / s), 0, L) (L = 255 for 8-bit, 15 for 4-bit
-// codes, one code per byte); 16 elements per thread per step.
+// codes, one code per byte).
 __device__ __forceinline__ uint32_t sq8_code(float x, float b, float s, float top) {
     float q = rintf(__fdiv_rn(__fsub_rn(x, b), s));
     q = (q >= 0.0f) ? q : 0.0f;
@@ -154,15 +154,45 @@ __device__ __forceinline__ uint32_t sq8_code(float x, float b, float s, float to
     return (uint32_t)q;
 }
 
+// The same code with one multiplication in place of the division: with
+// rs = fl(1/s) a normal number, q' = fl(a rs) (a = fl(x - b)) is within
+// (2^-23 + 2^-24 + 2^-48) |a/s| of the correctly rounded quotient q.  Only
+// quotients in [-0.5, L + 0.5] decide a code, and there |a/s| <= 256, so the two
+// are within 2^-14.4: when q' is more than 2^-13 away from every half-integer
+// they round to the same integer (quotients beyond that range clip to the same
+// end on both sides); otherwise (and for inf / NaN, including rs = NaN passed
+// for a subnormal 1/s) the quotient is taken by the IEEE division.
+__device__ __forceinline__ uint32_t sq8_code_rs(float x, float b, float s, float rs, float top) {
+    const float a = __fsub_rn(x, b);
+    const float q = __fmul_rn(a, rs);
+    float t = rintf(q);
+    if (!(fabsf(__fsub_rn(q, t)) < 0.5f - 0x1p-13f)) t = rintf(__fdiv_rn(a, s));
+    t = (t >= 0.0f) ? t : 0.0f;
+    t = fminf(t, top);
+    return (uint32_t)t;
+}
+
 // d % 4 == 0: one warp per row, lane l takes the float4 at dimensions
 // 128t + 4l .. + 3 and writes their four codes as one 32-bit word, so the
 // (b, s) loads and the code stores are contiguous across the warp; a row's
-// loads (up to SQ_V4 float4 per lane) are issued before use.
+// loads (up to SQ_V4 float4 per lane) are issued before use.  The block keeps
+// fl(1/s) per column in shared memory (sq8_code_rs).
 constexpr int SQ_V4 = 8;
+constexpr int SQ_RS_MAX_D = 8192;  // 32 KB of reciprocals
 
 __global__ void sq8_encode_rows_kernel(const float4 *__restrict__ X, int64_t n, int d,
                                        const float4 *__restrict__ b, const float4 *__restrict__ s,
                                        float top, uint32_t *__restrict__ out) {
+    extern __shared__ float4 sq_rs[];
+    for (int c = threadIdx.x; c < (d >> 2); c += blockDim.x) {
+        const float4 sv = __ldg(s + c);
+        auto rcp = [](float v) {
+            const float r = __frcp_rn(v);
+            return fabsf(r) >= 0x1p-126f ? r : __int_as_float(0x7fffffff);
+        };
+        sq_rs[c] = make_float4(rcp(sv.x), rcp(sv.y), rcp(sv.z), rcp(sv.w));
+    }
+    __syncthreads();
     const int lane = threadIdx.x & 31;
     const int64_t warp = (blockIdx.x * (int64_t)blockDim.x + threadIdx.x) >> 5;
     const int64_t nwarps = ((int64_t)gridDim.x * blockDim.x) >> 5;
@@ -181,9 +211,11 @@ __global__ void sq8_encode_rows_kernel(const float4 *__restrict__ X, int64_t n, 
             for (int u = 0; u < SQ_V4; ++u) {
                 const int j = 32 * (t0 + u) + lane;
                 if (j < d4) {
-                    const float4 bb = __ldg(b + j), ss = __ldg(s + j);
-                    o[j] = sq8_code(v[u].x, bb.x, ss.x, top) | (sq8_code(v[u].y, bb.y, ss.y, top) << 8) |
-                           (sq8_code(v[u].z, bb.z, ss.z, top) << 16) | (sq8_code(v[u].w, bb.w, ss.w, top) << 24);
+                    const float4 bb = __ldg(b + j), ss = __ldg(s + j), rr = sq_rs[j];
+                    o[j] = sq8_code_rs(v[u].x, bb.x, ss.x, rr.x, top) |
+                           (sq8_code_rs(v[u].y, bb.y, ss.y, rr.y, top) << 8) |
+                           (sq8_code_rs(v[u].z, bb.z, ss.z, rr.z, top) << 16) |
+                           (sq8_code_rs(v[u].w, bb.w, ss.w, rr.w, top) << 24);
                 }
             }
         }
@@ -212,8 +244,9 @@ cudaError_t launch_sq8_encode(const float *X, int64_t n, int d, const float *b, 
                               int levels, uint8_t *codes, cudaStream_t st) {
     const int64_t total = n * d;
     const float top = (float)levels;
-    if (d % 4 == 0 && (((uintptr_t)X | (uintptr_t)b | (uintptr_t)s) & 15) == 0 && ((uintptr_t)codes & 3) == 0) {
-        sq8_encode_rows_kernel<<<grid_for(n * 32, 256), 256, 0, st>>>(
+    if (d % 4 == 0 && d <= SQ_RS_MAX_D && (((uintptr_t)X | (uintptr_t)b | (uintptr_t)s) & 15) == 0 &&
+        ((uintptr_t)codes & 3) == 0) {
+        sq8_encode_rows_kernel<<<grid_for(n * 32, 256), 256, (size_t)d * sizeof(float), st>>>(
             reinterpret_cast<const float4 *>(X), n, d, reinterpret_cast<const float4 *>(b),
             reinterpret_cast<const float4 *>(s), top, reinterpret_cast<uint32_t *>(codes));
     } else {

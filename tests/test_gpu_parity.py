@@ -215,6 +215,33 @@ def test_quantize_sq8_bitexact(skm, n, d):
     np.testing.assert_array_equal(Y.cpu().numpy(), oracle.sq8_decode(q["codes"].cpu().numpy(), b, s))
 
 
+@pytest.mark.parametrize("bits", [8, 4])
+def test_quantize_sq8_half_integer_quotients(skm, bits):
+    """Fixed (b, s) per column, including scales whose reciprocal is subnormal or
+    infinite, and points whose quotients (x - b)/s sit at or one or two ulps
+    around every half-integer of the code range and beyond both ends."""
+    g = np.random.default_rng(bits)
+    d, n = 512, 600
+    L = 255 if bits == 8 else 15
+    b = g.uniform(-2, 2, size=d).astype(np.float32)
+    s = (g.uniform(0.01, 3, size=d) / L).astype(np.float32)
+    s[:4] = [1.0, 1.5 * 2.0 ** 127, 1e-40, 2.0 ** -126]
+    b[:4] = [0.0, 0.0, 0.0, 0.0]
+    m = g.integers(-4, 2 * L + 6, size=(n, d)).astype(np.float32) * np.float32(0.5)
+    with np.errstate(over="ignore", invalid="ignore"):
+        X = (b[None, :] + m * s[None, :]).astype(np.float32)
+    X[~np.isfinite(X)] = 0.0
+    nud = g.integers(-2, 3, size=(n, d))
+    for _k in range(2):
+        X = np.where(nud > 0, np.nextafter(X, np.float32(np.inf)), X)
+        X = np.where(nud < 0, np.nextafter(X, np.float32(-np.inf)), X)
+        nud = nud - np.sign(nud)
+    X = X.astype(np.float32)
+    q = skm.skm_quantize(skm.REPR_SQ8, torch.from_numpy(X).to(DEV), fit=False, b=torch.from_numpy(b).to(DEV),
+                         s=torch.from_numpy(s).to(DEV), bits=bits)
+    np.testing.assert_array_equal(q["codes"].cpu().numpy(), oracle.sq8_encode(X, b, s, bits=bits))
+
+
 @pytest.mark.parametrize("n,d,k", [(2000, 64, 50), (777, 33, 7), (1024, 1024, 129), (300, 5, 300),
                                    (600, 1500, 40), (1000, 1024, 1)])
 def test_assign_update_sq8_bitexact(skm, n, d, k):
@@ -738,6 +765,33 @@ def _lvq4_host(q, d):
                                  (257, 1020), (100, 1024)])
 def test_encode_lvq4_bitexact(skm, n, d):
     X = _points(n, d, seed=n + 3)
+    q = skm.skm_quantize(skm.REPR_LVQ4, X.to(DEV))
+    h = _lvq4_host(q, d)
+    codes, fac, _ = oracle.lvq4_encode(X.numpy())
+    np.testing.assert_array_equal(h["words"], oracle.lvq4_pack(codes))
+    np.testing.assert_array_equal(h["fac"], fac)
+
+
+@pytest.mark.parametrize("d", [768, 36])
+def test_encode_lvq4_half_integer_quotients(skm, d):
+    """Quotients (x - b)/s at, and one or two ulps around, every half-integer
+    0.5 .. 14.5 (where rounding half to even decides the code), with s = 1 and
+    with scales that are not powers of two."""
+    g = np.random.default_rng(d)
+    rows = []
+    for lo, span in [(0.0, 15.0), (-3.25, 1.5), (0.1, 15.0 * 0.37), (1e-3, 2.2e-3)]:
+        for _ in range(40):
+            s = np.float32(np.float32(span) / np.float32(15.0))
+            m = g.integers(0, 30, size=d).astype(np.float32) * np.float32(0.5)
+            x = (np.float32(lo) + m * s).astype(np.float32)
+            nud = g.integers(-2, 3, size=d)
+            for _k in range(2):
+                x = np.where(nud > 0, np.nextafter(x, np.float32(np.inf)), x)
+                x = np.where(nud < 0, np.nextafter(x, np.float32(-np.inf)), x)
+                nud = nud - np.sign(nud)
+            x[0], x[1] = np.float32(lo), np.float32(np.float32(lo) + np.float32(span))
+            rows.append(x.astype(np.float32))
+    X = torch.from_numpy(np.stack(rows))
     q = skm.skm_quantize(skm.REPR_LVQ4, X.to(DEV))
     h = _lvq4_host(q, d)
     codes, fac, _ = oracle.lvq4_encode(X.numpy())
