@@ -331,7 +331,10 @@ def run_ours(args):
         C_host32.copy_(C32)
         C_hostR.copy_(Cr)
         a_host = torch.empty(2, N_POINTS, dtype=torch.int32, pin_memory=True)
-        Xd2 = torch.empty_like(X)
+        # two device buffers for the points: step t + 1's copy streams in while
+        # step t is still being assigned and updated (the next step's points do
+        # not depend on this step; its centroids do, and wait for the D2H)
+        Xbuf = [torch.empty_like(X), torch.empty_like(X)]
         Cd32 = torch.empty_like(C32)
         CdR = torch.empty_like(Cr)
         # The H2D copy of the points is cut into E2E_CHUNKS row ranges on a copy
@@ -350,7 +353,7 @@ def run_ours(args):
         FE = torch.empty(N_POINTS, device=dev, dtype=torch.float32)
         popxE = torch.empty(N_POINTS, device=dev, dtype=torch.int32)
         mE = q["m"]
-        probe32 = skm.Points(skm.REPR_F32, Xd2[:cmax], DIM)
+        probe32 = skm.Points(skm.REPR_F32, Xbuf[0][:cmax], DIM)
         wsA2 = skm.workspace(skm.OP_ASSIGN, probe32, K)
         wsAR2 = skm.workspace(skm.OP_ASSIGN, skm.Points(skm.REPR_RBQ1, codesE[:cmax], DIM, nx2E[:cmax],
                                                         FE[:cmax], popxE[:cmax], mE, e), K)
@@ -358,66 +361,92 @@ def run_ours(args):
         part32e = torch.zeros(K, DIM, device=dev, dtype=torch.float64)
         cnt32e = torch.zeros(K, device=dev, dtype=torch.int64)
         wsU2 = skm.workspace(skm.OP_UPDATE, probe32, K)
-        copy_stream = torch.cuda.Stream()
-        landed = [torch.cuda.Event() for _ in range(nchunk)]
+        copy_stream = torch.cuda.Stream()   # the points, one step ahead
+        cent_stream = torch.cuda.Stream()   # the centroids, after the previous step's D2H
+        e2e_steps = max(2, min(args.steps, 5))
+        landed = [[torch.cuda.Event() for _ in range(nchunk)] for _ in range(2)]
         c_landed = torch.cuda.Event()
+        buf_free = [torch.cuda.Event(), torch.cuda.Event()]
+        d2h_done = torch.cuda.Event()
         # per-range point descriptors over the fixed device buffers (views)
-        pcs = [skm.Points(skm.REPR_F32, Xd2[b0:b1], DIM) for b0, b1 in bounds]
+        pcs = [[skm.Points(skm.REPR_F32, xb[b0:b1], DIM) for b0, b1 in bounds] for xb in Xbuf]
         qouts = [{"codes": codesE[b0:b1], "nx2": nx2E[b0:b1], "F": FE[b0:b1], "popx": popxE[b0:b1]}
                  for b0, b1 in bounds]
         prcs = [skm.Points(skm.REPR_RBQ1, codesE[b0:b1], DIM, nx2E[b0:b1], FE[b0:b1], popxE[b0:b1], mE, e)
                 for b0, b1 in bounds]
-        pall = skm.Points(skm.REPR_F32, Xd2, DIM)
+        pall = [skm.Points(skm.REPR_F32, xb, DIM) for xb in Xbuf]
         host_ms = []
         h2d = X_host.numel() * 4 + 2 * K * DIM * 4
         d2h = 2 * N_POINTS * 4 + 2 * K * DIM * 4
-        e2e_steps = max(2, min(args.steps, 5))
         # the host link's copy rate just before the run (the e2e step is bound by
         # it; it varies with other traffic on the shared host)
         torch.cuda.synchronize()
         p0, p1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
         p0.record(stream)
-        Xd2.copy_(X_host, non_blocking=True)
+        Xbuf[0].copy_(X_host, non_blocking=True)
         p1.record(stream)
         torch.cuda.synchronize()
         h2d_probe_gbs = X_host.numel() * 4 / (p0.elapsed_time(p1) / 1e3) / 1e9
+
+        def enqueue_points(t):
+            slot = t % 2
+            if t >= 2:
+                copy_stream.wait_event(buf_free[slot])  # step t - 2 is done with this buffer
+            with torch.cuda.stream(copy_stream):
+                for (b0, b1), ev in zip(bounds, landed[slot]):
+                    Xbuf[slot][b0:b1].copy_(X_host[b0:b1], non_blocking=True)
+                    ev.record(copy_stream)
+
+        def e2e_run(nsteps):
+            """nsteps end-to-end steps; the device time from the first copy to the
+            last step's D2H (ms)."""
+            s0, s1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            s0.record(stream)
+            copy_stream.wait_stream(stream)
+            cent_stream.wait_stream(stream)
+            enqueue_points(0)
+            for t in range(nsteps):
+                th0 = time.perf_counter()
+                slot = t % 2
+                if t + 1 < nsteps:
+                    enqueue_points(t + 1)
+                if t > 0:
+                    cent_stream.wait_event(d2h_done)  # this step's centroids are the last step's results
+                # by the SMs, not a copy engine: there they would queue behind the
+                # next step's point ranges
+                skm.skm_copy_from_host(Cd32, C_host32, stream=cent_stream)
+                skm.skm_copy_from_host(CdR, C_hostR, stream=cent_stream)
+                c_landed.record(cent_stream)
+                stream.wait_event(c_landed)
+                part32e.zero_()
+                cnt32e.zero_()
+                xb = Xbuf[slot]
+                for (b0, b1), ev, pc, qo, prc in zip(bounds, landed[slot], pcs[slot], qouts, prcs):
+                    stream.wait_event(ev)
+                    skm.skm_assign(pc, Cd32, K, want_dist=False, ws=wsA2, out=a32[b0:b1])
+                    skm.skm_update(pc, a32[b0:b1], None, counts=cnt32e, partial=part32e, ws=wsU2)
+                    skm.skm_quantize(skm.REPR_RBQ1, xb[b0:b1], fit=False, m=mE, ws=wsQ2, out=qo)
+                    skm.skm_assign(prc, CdR, K, want_dist=False, ws=wsAR2, out=aR[b0:b1])
+                buf_free[slot].record(stream)
+                skm.skm_update_finalize(pall[slot], part32e, cnt32e, Cd32)
+                host_ms.append((time.perf_counter() - th0) * 1e3)  # enqueue only (no sync so far)
+                eE = skm.skm_rbq1_exponent(FE)
+                pR2 = skm.Points(skm.REPR_RBQ1, codesE, DIM, nx2E, FE, popxE, mE, eE)
+                skm.skm_update(pR2, aR, CdR, counts=cntR, ws=wsUR)
+                a_host[0].copy_(a32, non_blocking=True)
+                a_host[1].copy_(aR, non_blocking=True)
+                C_host32.copy_(Cd32, non_blocking=True)
+                C_hostR.copy_(CdR, non_blocking=True)
+                d2h_done.record(stream)
+            s1.record(stream)
+            torch.cuda.synchronize()
+            return s0.elapsed_time(s1)
+
+        e2e_run(2)  # warm-up (first-use costs of the range-sized calls), untimed
+        host_ms.clear()
         if world > 1:
             dist.barrier()
-        s0, s1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-        s0.record(stream)
-        for _ in range(e2e_steps):
-            th0 = time.perf_counter()
-            copy_stream.wait_stream(stream)  # the previous step is done with Xd2 and the centroids
-            with torch.cuda.stream(copy_stream):
-                # centroids first: queued behind the point ranges on the same copy
-                # engine they would hold back every range's work
-                Cd32.copy_(C_host32, non_blocking=True)
-                CdR.copy_(C_hostR, non_blocking=True)
-                c_landed.record(copy_stream)
-                for (b0, b1), ev in zip(bounds, landed):
-                    Xd2[b0:b1].copy_(X_host[b0:b1], non_blocking=True)
-                    ev.record(copy_stream)
-            stream.wait_event(c_landed)
-            part32e.zero_()
-            cnt32e.zero_()
-            for (b0, b1), ev, pc, qo, prc in zip(bounds, landed, pcs, qouts, prcs):
-                stream.wait_event(ev)
-                skm.skm_assign(pc, Cd32, K, want_dist=False, ws=wsA2, out=a32[b0:b1])
-                skm.skm_update(pc, a32[b0:b1], None, counts=cnt32e, partial=part32e, ws=wsU2)
-                skm.skm_quantize(skm.REPR_RBQ1, Xd2[b0:b1], fit=False, m=mE, ws=wsQ2, out=qo)
-                skm.skm_assign(prc, CdR, K, want_dist=False, ws=wsAR2, out=aR[b0:b1])
-            skm.skm_update_finalize(pall, part32e, cnt32e, Cd32)
-            host_ms.append((time.perf_counter() - th0) * 1e3)  # enqueue only (no sync so far)
-            eE = skm.skm_rbq1_exponent(FE)
-            pR2 = skm.Points(skm.REPR_RBQ1, codesE, DIM, nx2E, FE, popxE, mE, eE)
-            skm.skm_update(pR2, aR, CdR, counts=cntR, ws=wsUR)
-            a_host[0].copy_(a32, non_blocking=True)
-            a_host[1].copy_(aR, non_blocking=True)
-            C_host32.copy_(Cd32, non_blocking=True)
-            C_hostR.copy_(CdR, non_blocking=True)
-        s1.record(stream)
-        torch.cuda.synchronize()
-        ems = s0.elapsed_time(s1)
+        ems = e2e_run(e2e_steps)
         if world > 1:
             t = torch.tensor([ems], device=dev, dtype=torch.float64)
             dist.all_reduce(t, op=dist.ReduceOp.MAX)
@@ -427,9 +456,10 @@ def run_ours(args):
                "host_enqueue_ms_per_step": round(statistics.mean(host_ms), 3),
                "h2d_probe_gbs": round(h2d_probe_gbs, 1),
                "ms_per_step": ems / e2e_steps,
-               "path": f"pinned host fp32 points -> H2D in {nchunk} row ranges on a copy stream, each "
-                       "range assigned (fp32) and encoded + assigned (1-bit) once it has landed -> "
-                       "skm_update (fp32, 1-bit) -> D2H assignments + centroids"}
+               "path": f"pinned host fp32 points -> H2D in {nchunk} row ranges on a copy stream (two device "
+                       "buffers: the next step's points stream in during this step's tail), each range assigned "
+                       "(fp32) and encoded + assigned (1-bit) once it has landed -> skm_update (fp32, 1-bit) -> "
+                       "D2H assignments + centroids, which the next step copies back as its centroids"}
 
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:

@@ -168,6 +168,19 @@ int skm_project(const float *X, int64_t n, int d, const float *mean, const float
 int skm_unproject(const float *Y, int64_t n, int d_out, const float *P, const float *mean, int d,
                   float *X, void *stream);
 
+/* Host-to-device copy by the SMs: bytes bytes from src_host (host memory the
+ * device can address: page-locked memory mapped into the device address space,
+ * e.g. cudaHostAlloc or a pinned PyTorch tensor; on hardware-coherent host
+ * links any host memory) to dst (device), loaded over the host link by a small
+ * grid of thread blocks instead of a copy engine.  A copy-engine copy can wait
+ * behind larger copies queued before it on the same engine; this call lets a
+ * small input (a step's centroids) land while a large one (the next step's
+ * points) is still streaming in.  The device address of src_host comes from
+ * cudaHostGetDevicePointer: when that fails the call returns
+ * SKM_ERR_INVALID_ARG and launches nothing.  bytes = 0 is a no-op.
+ * Asynchronous on stream: src_host must stay valid until the copy is done. */
+int skm_copy_from_host(void *dst, const void *src_host, size_t bytes, void *stream);
+
 /* Randomized Hadamard rotation (a structured random orthogonal transform in
  * place of a dense random rotation before RabitQ / SuperKMeans, Section 3.1;
  * O(D log D) per point): Y = (1/sqrt(D)) H_D diag(sigma) [X - mean; 0] with

@@ -35,7 +35,8 @@ _lib = None
 # Every entry point declared in include/skm.h.
 EXPORTED_SYMBOLS = [
     "skm_last_error", "skm_version", "skm_kernel_launches", "skm_workspace_size", "skm_screen_bytes",
-    "skm_screen_prep", "skm_project", "skm_project_hadamard", "skm_unproject", "skm_make_rotation",
+    "skm_screen_prep", "skm_project", "skm_project_hadamard", "skm_unproject", "skm_copy_from_host",
+    "skm_make_rotation",
     "skm_pca_fit", "skm_quantize", "skm_rbq1_exponent", "skm_lvq4_exponent", "skm_assign", "skm_assign_rbq1_noalloc",
     "skm_assign_segmented",
     "skm_update",
@@ -108,6 +109,7 @@ def lib():
             "skm_make_rotation": ([u64, i32, vp], i32),
             "skm_project_hadamard": ([vp, i64, i32, vp, vp, i32, i32, vp, vp], i32),
             "skm_unproject": ([vp, i64, i32, vp, vp, i32, vp, vp], i32),
+            "skm_copy_from_host": ([vp, vp, sz, vp], i32),
             "skm_pca_fit": ([vp, i64, i32, i32, vp, vp, vp, vp, sz, vp], i32),
             "skm_quantize": ([i32, vp, i64, i32, vp, vp, vp, sz, vp], i32),
             "skm_rbq1_exponent": ([vp, i64, vp, vp, sz, vp], i32),
@@ -239,6 +241,16 @@ def skm_project_hadamard(X, sigma, mean=None, out_dtype=DTYPE_F32, stream=None):
     _check(lib().skm_project_hadamard(_ptr(X), n, d, _ptr(mean), _ptr(sigma), int(D), out_dtype, _ptr(Y),
                                       _stream(stream)))
     return Y
+
+
+def skm_copy_from_host(dst, src, stream=None):
+    """dst (contiguous device tensor) <- src (contiguous pinned host tensor of
+    the same number of bytes), copied by thread blocks over the host link."""
+    nb = src.numel() * src.element_size()
+    if not dst.is_contiguous() or not src.is_contiguous() or dst.numel() * dst.element_size() != nb:
+        raise ValueError("skm_copy_from_host: contiguous tensors of equal byte size")
+    _check(lib().skm_copy_from_host(_ptr(dst), _ptr(src), nb, _stream(stream)))
+    return dst
 
 
 def skm_unproject(Y, P, mean=None, stream=None):

@@ -491,4 +491,36 @@ cudaError_t launch_unproject(const float *Y, int64_t n, int dout, const float *P
     return launched();
 }
 
+// Host-to-device copy by the SMs (skm_copy_from_host): 16-byte loads from the
+// mapped host buffer, four in flight per thread, when both ends are 16-byte
+// aligned; bytes otherwise and for the tail.  A few dozen blocks fill the host
+// link.
+__global__ void copy_from_host_kernel(const uint8_t *__restrict__ src, uint8_t *__restrict__ dst, size_t bytes,
+                                      size_t n16) {
+    const size_t stride = (size_t)gridDim.x * blockDim.x;
+    size_t i = blockIdx.x * (size_t)blockDim.x + threadIdx.x;
+    const uint4 *s4 = reinterpret_cast<const uint4 *>(src);
+    uint4 *d4 = reinterpret_cast<uint4 *>(dst);
+    for (; i + 3 * stride < n16; i += 4 * stride) {
+        const uint4 a = s4[i], b = s4[i + stride], c = s4[i + 2 * stride], e = s4[i + 3 * stride];
+        d4[i] = a;
+        d4[i + stride] = b;
+        d4[i + 2 * stride] = c;
+        d4[i + 3 * stride] = e;
+    }
+    for (; i < n16; i += stride) d4[i] = s4[i];
+    for (size_t j = 16 * n16 + blockIdx.x * (size_t)blockDim.x + threadIdx.x; j < bytes; j += stride) dst[j] = src[j];
+}
+
+cudaError_t launch_copy_from_host(const void *src, void *dst, size_t bytes, cudaStream_t st) {
+    if (bytes == 0) return cudaSuccess;
+    const bool al = (((uintptr_t)src | (uintptr_t)dst) & 15) == 0;
+    const size_t n16 = al ? bytes / 16 : 0;
+    const size_t units = al ? n16 : bytes;
+    const size_t blocks = (units + 255) / 256;
+    copy_from_host_kernel<<<(unsigned)(blocks < 32 ? (blocks < 1 ? 1 : blocks) : 32), 256, 0, st>>>(
+        static_cast<const uint8_t *>(src), static_cast<uint8_t *>(dst), bytes, n16);
+    return launched();
+}
+
 }  // namespace skm

@@ -454,6 +454,20 @@ int skm_unproject(const float *Y, int64_t n, int d_out, const float *P, const fl
     return SKM_OK;
 }
 
+int skm_copy_from_host(void *dst, const void *src_host, size_t bytes, void *stream) {
+    if (bytes == 0) return SKM_OK;
+    if (!dst || !src_host) return set_error(SKM_ERR_INVALID_ARG, "NULL pointer");
+    void *src_dev = nullptr;
+    const cudaError_t e = cudaHostGetDevicePointer(&src_dev, const_cast<void *>(src_host), 0);
+    if (e != cudaSuccess || !src_dev) {
+        (void)cudaGetLastError();  // clear the failed query's (non-sticky) error
+        return set_error(SKM_ERR_INVALID_ARG, "src_host is not mapped page-locked host memory (%s)",
+                         cudaGetErrorString(e));
+    }
+    SKM_CUDA_TRY(launch_copy_from_host(src_dev, dst, bytes, S(stream)));
+    return SKM_OK;
+}
+
 int skm_make_rotation(uint64_t seed, int d, float *P_host) {
     if (!P_host || d < 1 || d > MAX_D) return set_error(SKM_ERR_INVALID_ARG, "bad arguments");
     std::vector<double> A((size_t)d * d);

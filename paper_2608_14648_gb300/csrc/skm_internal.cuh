@@ -239,6 +239,8 @@ cudaError_t launch_cov_reduce(const double *partial, int splits, int d, double *
 
 // LVQ4 (Section 3.1 "LVQ4"; k_lvq4.cu).  Codes: uint32 [n][ceil(d/8)] nibbles;
 // per-vector terms float4 (s, b, N, A) for points, (s, b, N, G) for centroids.
+// dst (device) <- src (device address of mapped page-locked host memory)
+cudaError_t launch_copy_from_host(const void *src, void *dst, size_t bytes, cudaStream_t st);
 __host__ __device__ inline int lvq4_words(int d) { return (d + 7) / 8; }
 cudaError_t launch_lvq4_encode(const float *X, int64_t n, int d, uint32_t *codes, float4 *fac,
                                cudaStream_t st);

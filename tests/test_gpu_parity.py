@@ -710,6 +710,38 @@ def test_fit_hierarchical_f32_vs_oracle(skm):
     assert abs(wg - wo) / wo <= 1e-3
 
 
+# ------------------------------------------- host-to-device copy by the SMs
+@pytest.mark.parametrize("nbytes,offset", [(6 * 1024 * 1024 + 48, 0), (1000003, 3), (15, 1), (16, 0)])
+def test_copy_from_host(skm, nbytes, offset):
+    g = torch.Generator().manual_seed(nbytes)
+    src_all = torch.randint(0, 256, (nbytes + offset,), dtype=torch.uint8, generator=g).pin_memory()
+    src = src_all[offset:]
+    dst_all = torch.zeros(nbytes + 1, dtype=torch.uint8, device=DEV)
+    dst = dst_all[1:] if offset else dst_all[:nbytes]
+    skm.skm_copy_from_host(dst, src)
+    torch.cuda.synchronize()
+    assert torch.equal(dst.cpu(), src)
+    # the guard byte outside the destination is untouched
+    assert int(dst_all[0 if offset else nbytes].item()) == 0
+
+
+def test_copy_from_host_pageable_memory(skm):
+    """Ordinary (pageable) host memory: copied where the device addresses all
+    host memory (a hardware-coherent host link), else refused before any launch."""
+    src = torch.arange(4096, dtype=torch.float32)
+    dst = torch.zeros(4096, dtype=torch.float32, device=DEV)
+    try:
+        skm.skm_copy_from_host(dst, src)
+        refused = False
+    except skm.SkmError:
+        refused = True
+    torch.cuda.synchronize()
+    if refused:
+        assert float(dst.abs().sum().item()) == 0.0
+    else:
+        assert torch.equal(dst.cpu(), src)
+
+
 # ------------------------------------- centroids back in the original space
 @pytest.mark.parametrize("k,d,dout", [(300, 96, 32), (1000, 1024, 256), (17, 50, 50)])
 def test_unproject_vs_oracle(skm, k, d, dout):
