@@ -138,11 +138,10 @@ __global__ void lvq4_encode_kernel(const float *__restrict__ X, int64_t n, int d
 }
 
 // d % 4 == 0 and d <= 1024: the row stays in registers (lane l holds the
-// float4 at dimensions 128u + 4l .. + 3, all loads issued at once), so the
-// points are read once; the two lanes of a pair assemble one nibble word
-// (8 dimensions), the even lane stores it.  Same code arithmetic as
-// lvq4_encode_warp.
-constexpr int LVQ_V4 = 8;
+// float4 at dimensions 128u + 4l .. + 3 for u < NV = ceil(d / 128), the next
+// row's loads in flight while this one is encoded), so the points are read
+// once; the two lanes of a pair assemble one nibble word (8 dimensions), the
+// even lane stores it.  Same code arithmetic as lvq4_encode_warp.
 
 // clip(rint(fl((x - lo) / s)), 0, 15) with one multiplication in place of the
 // division: with rs = fl(1/s), q' = fl(a rs) (a = fl(x - lo)) is within
@@ -152,34 +151,55 @@ constexpr int LVQ_V4 = 8;
 // 2^-17 away from every half-integer, q and q' round to the same integer;
 // otherwise (and for inf / NaN) the quotient is taken by the IEEE division.
 // The bound needs a normal rs: callers pass NaN instead of a subnormal one.
-__device__ __forceinline__ uint32_t lvq4_code(float x, float lo, float s, float rs) {
-    const float a = __fsub_rn(x, lo);
-    float q = __fmul_rn(a, rs);
-    float t = rintf(q);
-    if (!(fabsf(__fsub_rn(q, t)) < 0.5f - 0x1p-17f)) t = rintf(__fdiv_rn(a, s));
-    t = (t >= 0.0f) ? t : 0.0f;
-    t = fminf(t, 15.0f);
-    return (uint32_t)t;
+// Four codes at once: one combined test sends the float4 to the divisions
+// when any of its quotients is near a half-integer or not finite (fmaxf drops
+// NaN, hence the separate finiteness test).
+__device__ __forceinline__ void lvq4_code4(const float4 &x, float lo, float s, float rs, uint32_t &c0, uint32_t &c1,
+                                           uint32_t &c2, uint32_t &c3) {
+    const float ax = __fsub_rn(x.x, lo), ay = __fsub_rn(x.y, lo), az = __fsub_rn(x.z, lo), aw = __fsub_rn(x.w, lo);
+    const float qx = __fmul_rn(ax, rs), qy = __fmul_rn(ay, rs), qz = __fmul_rn(az, rs), qw = __fmul_rn(aw, rs);
+    float tx = rintf(qx), ty = rintf(qy), tz = rintf(qz), tw = rintf(qw);
+    constexpr float lim = 0.5f - 0x1p-17f;
+    if (!(fmaxf(fmaxf(fabsf(__fsub_rn(qx, tx)), fabsf(__fsub_rn(qy, ty))),
+                fmaxf(fabsf(__fsub_rn(qz, tz)), fabsf(__fsub_rn(qw, tw)))) < lim) ||
+        !(fabsf(qx) + fabsf(qy) + fabsf(qz) + fabsf(qw) < INFINITY)) {
+        if (!(fabsf(__fsub_rn(qx, tx)) < lim)) tx = rintf(__fdiv_rn(ax, s));
+        if (!(fabsf(__fsub_rn(qy, ty)) < lim)) ty = rintf(__fdiv_rn(ay, s));
+        if (!(fabsf(__fsub_rn(qz, tz)) < lim)) tz = rintf(__fdiv_rn(az, s));
+        if (!(fabsf(__fsub_rn(qw, tw)) < lim)) tw = rintf(__fdiv_rn(aw, s));
+    }
+    auto clip = [](float t) { return (uint32_t)fminf(t >= 0.0f ? t : 0.0f, 15.0f); };
+    c0 = clip(tx);
+    c1 = clip(ty);
+    c2 = clip(tz);
+    c3 = clip(tw);
 }
 
-__global__ void __launch_bounds__(256, 3) lvq4_encode_v4_kernel(const float4 *__restrict__ X, int64_t n, int d, uint32_t *__restrict__ codes,
-                                      float4 *__restrict__ fac) {
+
+template <int NV>
+__global__ void __launch_bounds__(256, 2) lvq4_encode_v4_kernel(const float4 *__restrict__ X, int64_t n, int d,
+                                                                uint32_t *__restrict__ codes, float4 *__restrict__ fac) {
     const int lane = threadIdx.x & 31;
     const int64_t w0 = (blockIdx.x * (int64_t)blockDim.x + threadIdx.x) >> 5;
     const int64_t nw = ((int64_t)gridDim.x * blockDim.x) >> 5;
     const int W = lvq4_words(d), d4 = d >> 2;
-    FacBatch fb;
-    for (int64_t p = w0; p < n; p += nw) {
+    auto load_row = [&](int64_t p, float4(&v)[NV]) {
         const float4 *x = X + p * d4;
-        float4 v[LVQ_V4];
-        float lo = INFINITY, hi = -INFINITY;
 #pragma unroll
-        for (int u = 0; u < LVQ_V4; ++u) {
+        for (int u = 0; u < NV; ++u) {
             const int j = 32 * u + lane;
             if (j < d4) v[u] = __ldg(x + j);
         }
+    };
+    FacBatch fb;
+    float4 v[NV];
+    if (w0 < n) load_row(w0, v);
+    for (int64_t p = w0; p < n; p += nw) {
+        float4 nxt[NV];
+        if (p + nw < n) load_row(p + nw, nxt);  // the next row in flight while this one is encoded
+        float lo = INFINITY, hi = -INFINITY;
 #pragma unroll
-        for (int u = 0; u < LVQ_V4; ++u) {
+        for (int u = 0; u < NV; ++u) {
             if (32 * u + lane < d4) {
                 lo = fminf(lo, fminf(fminf(v[u].x, v[u].y), fminf(v[u].z, v[u].w)));
                 hi = fmaxf(hi, fmaxf(fmaxf(v[u].x, v[u].y), fmaxf(v[u].z, v[u].w)));
@@ -197,25 +217,25 @@ __global__ void __launch_bounds__(256, 3) lvq4_encode_v4_kernel(const float4 *__
         int32_t S = 0, Q = 0;
         uint32_t *cw = codes + p * W;
 #pragma unroll
-        for (int u = 0; u < LVQ_V4; ++u) {
-            if (32 * u < d4) {  // warp-uniform
-                const int j = 32 * u + lane;
-                uint32_t h = 0;
-                if (j < d4) {
-                    const uint32_t c0 = lvq4_code(v[u].x, lo, s, rs), c1 = lvq4_code(v[u].y, lo, s, rs);
-                    const uint32_t c2 = lvq4_code(v[u].z, lo, s, rs), c3 = lvq4_code(v[u].w, lo, s, rs);
-                    S += (int32_t)(c0 + c1 + c2 + c3);
-                    Q += (int32_t)(c0 * c0 + c1 * c1 + c2 * c2 + c3 * c3);
-                    h = (c0 | (c1 << 4) | (c2 << 8) | (c3 << 12)) << (16 * (lane & 1));
-                }
-                h |= __shfl_xor_sync(FULL, h, 1);
-                const int wi = j >> 1;
-                if ((lane & 1) == 0 && wi < W) cw[wi] = h;
+        for (int u = 0; u < NV; ++u) {
+            const int j = 32 * u + lane;
+            uint32_t h = 0;
+            if (j < d4) {
+                uint32_t c0, c1, c2, c3;
+                lvq4_code4(v[u], lo, s, rs, c0, c1, c2, c3);
+                S += (int32_t)(c0 + c1 + c2 + c3);
+                Q += (int32_t)(c0 * c0 + c1 * c1 + c2 * c2 + c3 * c3);
+                h = (c0 | (c1 << 4) | (c2 << 8) | (c3 << 12)) << (16 * (lane & 1));
             }
+            h |= __shfl_xor_sync(FULL, h, 1);
+            const int wi = j >> 1;
+            if ((lane & 1) == 0 && wi < W) cw[wi] = h;
         }
         S = __reduce_add_sync(FULL, S);
         Q = __reduce_add_sync(FULL, Q);
         fb.put(Lvq4Vec{lo, s, S, Q}, p, lane, fac, d);
+#pragma unroll
+        for (int u = 0; u < NV; ++u) v[u] = nxt[u];
     }
     fb.flush(fac, d);
 }
@@ -477,11 +497,22 @@ __global__ void lvq4_decode_rows_kernel(const uint32_t *__restrict__ codes, cons
 }  // namespace
 
 cudaError_t launch_lvq4_encode(const float *X, int64_t n, int d, uint32_t *codes, float4 *fac, cudaStream_t st) {
-    if (d % 4 == 0 && d <= 32 * 4 * LVQ_V4 && ((uintptr_t)X & 15) == 0)
-        lvq4_encode_v4_kernel<<<grid_warps_rows(n), 256, 0, st>>>(reinterpret_cast<const float4 *>(X), n, d, codes,
-                                                                   fac);
-    else
-        lvq4_encode_kernel<<<grid_warps_rows(n), 256, 0, st>>>(X, n, d, codes, fac);
+    const float4 *X4 = reinterpret_cast<const float4 *>(X);
+    const int g = grid_warps_rows(n);
+    if (d % 4 == 0 && d <= 1024 && ((uintptr_t)X & 15) == 0) {
+        switch ((d + 127) / 128) {
+        case 1: lvq4_encode_v4_kernel<1><<<g, 256, 0, st>>>(X4, n, d, codes, fac); break;
+        case 2: lvq4_encode_v4_kernel<2><<<g, 256, 0, st>>>(X4, n, d, codes, fac); break;
+        case 3: lvq4_encode_v4_kernel<3><<<g, 256, 0, st>>>(X4, n, d, codes, fac); break;
+        case 4: lvq4_encode_v4_kernel<4><<<g, 256, 0, st>>>(X4, n, d, codes, fac); break;
+        case 5: lvq4_encode_v4_kernel<5><<<g, 256, 0, st>>>(X4, n, d, codes, fac); break;
+        case 6: lvq4_encode_v4_kernel<6><<<g, 256, 0, st>>>(X4, n, d, codes, fac); break;
+        case 7: lvq4_encode_v4_kernel<7><<<g, 256, 0, st>>>(X4, n, d, codes, fac); break;
+        default: lvq4_encode_v4_kernel<8><<<g, 256, 0, st>>>(X4, n, d, codes, fac); break;
+        }
+    } else {
+        lvq4_encode_kernel<<<g, 256, 0, st>>>(X, n, d, codes, fac);
+    }
     return launched();
 }
 

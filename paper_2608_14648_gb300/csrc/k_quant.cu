@@ -6,6 +6,15 @@
 
 namespace skm {
 
+static int grid_for(int64_t work, int threads) {
+    int64_t g = (work + threads - 1) / threads;
+    const int64_t cap = 152LL * 16;  // grid-stride kernels: at most 16 blocks per SM of 152
+    if (g > cap) g = cap;
+    if (g < 1) g = 1;
+    return (int)g;
+}
+
+
 // ---------------------------------------------------------------------------
 // Column min/max and column sums: blocks take a contiguous slab of rows; each
 // thread owns columns (strided by blockDim.x).  Partial results per slab are
@@ -222,6 +231,80 @@ __global__ void sq8_encode_rows_kernel(const float4 *__restrict__ X, int64_t n, 
     }
 }
 
+// d % 4 == 0 and d <= 1024: the layout of sq8_encode_rows_kernel with
+// NV = ceil(d / 128) float4 per lane and the next row's loads in flight while
+// the current row is coded.
+template <int NV>
+__global__ void __launch_bounds__(256) sq8_encode_pf_kernel(const float4 *__restrict__ X, int64_t n, int d,
+                                                            const float4 *__restrict__ b,
+                                                            const float4 *__restrict__ s, float top,
+                                                            uint32_t *__restrict__ out) {
+    __shared__ float4 rs_sh[256];
+    for (int c = threadIdx.x; c < (d >> 2); c += blockDim.x) {
+        const float4 sv = __ldg(s + c);
+        auto rcp = [](float v) {
+            const float r = __frcp_rn(v);
+            return fabsf(r) >= 0x1p-126f ? r : __int_as_float(0x7fffffff);
+        };
+        rs_sh[c] = make_float4(rcp(sv.x), rcp(sv.y), rcp(sv.z), rcp(sv.w));
+    }
+    __syncthreads();
+    const int lane = threadIdx.x & 31;
+    const int64_t warp = (blockIdx.x * (int64_t)blockDim.x + threadIdx.x) >> 5;
+    const int64_t nwarps = ((int64_t)gridDim.x * blockDim.x) >> 5;
+    const int d4 = d >> 2;
+    auto load_row = [&](int64_t p, float4(&v)[NV]) {
+        const float4 *x = X + p * d4;
+#pragma unroll
+        for (int u = 0; u < NV; ++u) {
+            const int j = 32 * u + lane;
+            if (j < d4) v[u] = __ldg(x + j);
+        }
+    };
+    float4 v[NV];
+    if (warp < n) load_row(warp, v);
+    for (int64_t p = warp; p < n; p += nwarps) {
+        float4 nxt[NV];
+        if (p + nwarps < n) load_row(p + nwarps, nxt);
+        uint32_t *o = out + p * d4;
+#pragma unroll
+        for (int u = 0; u < NV; ++u) {
+            const int j = 32 * u + lane;
+            if (j < d4) {
+                const float4 bb = __ldg(b + j), rr = rs_sh[j];
+                const float ax = __fsub_rn(v[u].x, bb.x), ay = __fsub_rn(v[u].y, bb.y);
+                const float az = __fsub_rn(v[u].z, bb.z), aw = __fsub_rn(v[u].w, bb.w);
+                const float qx = __fmul_rn(ax, rr.x), qy = __fmul_rn(ay, rr.y);
+                const float qz = __fmul_rn(az, rr.z), qw = __fmul_rn(aw, rr.w);
+                float tx = rintf(qx), ty = rintf(qy), tz = rintf(qz), tw = rintf(qw);
+                // any quotient near a half-integer (or not finite): the divisions decide
+                constexpr float lim = 0.5f - 0x1p-13f;
+                if (!(fmaxf(fmaxf(fabsf(__fsub_rn(qx, tx)), fabsf(__fsub_rn(qy, ty))),
+                            fmaxf(fabsf(__fsub_rn(qz, tz)), fabsf(__fsub_rn(qw, tw)))) < lim) ||
+                    !(fabsf(qx) + fabsf(qy) + fabsf(qz) + fabsf(qw) < INFINITY)) {
+                    const float4 ss = __ldg(s + j);
+                    if (!(fabsf(__fsub_rn(qx, tx)) < lim)) tx = rintf(__fdiv_rn(ax, ss.x));
+                    if (!(fabsf(__fsub_rn(qy, ty)) < lim)) ty = rintf(__fdiv_rn(ay, ss.y));
+                    if (!(fabsf(__fsub_rn(qz, tz)) < lim)) tz = rintf(__fdiv_rn(az, ss.z));
+                    if (!(fabsf(__fsub_rn(qw, tw)) < lim)) tw = rintf(__fdiv_rn(aw, ss.w));
+                }
+                auto clip = [top](float t) { return (uint32_t)fminf(t >= 0.0f ? t : 0.0f, top); };
+                o[j] = clip(tx) | (clip(ty) << 8) | (clip(tz) << 16) | (clip(tw) << 24);
+            }
+        }
+#pragma unroll
+        for (int u = 0; u < NV; ++u) v[u] = nxt[u];
+    }
+}
+
+template <int NV>
+static void sq8_pf_launch(const float *X, int64_t n, int d, const float *b, const float *s, float top,
+                          uint8_t *codes, cudaStream_t st) {
+    sq8_encode_pf_kernel<NV><<<grid_for(n * 32, 256), 256, 0, st>>>(
+        reinterpret_cast<const float4 *>(X), n, d, reinterpret_cast<const float4 *>(b),
+        reinterpret_cast<const float4 *>(s), top, reinterpret_cast<uint32_t *>(codes));
+}
+
 __global__ void sq8_encode_scalar_kernel(const float *__restrict__ X, int64_t total, int d,
                                          const float *__restrict__ b, const float *__restrict__ s,
                                          float top, uint8_t *__restrict__ out) {
@@ -232,20 +315,24 @@ __global__ void sq8_encode_scalar_kernel(const float *__restrict__ X, int64_t to
     }
 }
 
-static int grid_for(int64_t work, int threads) {
-    int64_t g = (work + threads - 1) / threads;
-    const int64_t cap = 152LL * 16;  // 16 resident blocks per SM on 152 SMs
-    if (g > cap) g = cap;
-    if (g < 1) g = 1;
-    return (int)g;
-}
-
 cudaError_t launch_sq8_encode(const float *X, int64_t n, int d, const float *b, const float *s,
                               int levels, uint8_t *codes, cudaStream_t st) {
     const int64_t total = n * d;
     const float top = (float)levels;
-    if (d % 4 == 0 && d <= SQ_RS_MAX_D && (((uintptr_t)X | (uintptr_t)b | (uintptr_t)s) & 15) == 0 &&
-        ((uintptr_t)codes & 3) == 0) {
+    const bool v4 = d % 4 == 0 && (((uintptr_t)X | (uintptr_t)b | (uintptr_t)s) & 15) == 0 &&
+                    ((uintptr_t)codes & 3) == 0;
+    if (v4 && d <= 1024) {
+        switch ((d + 127) / 128) {
+        case 1: sq8_pf_launch<1>(X, n, d, b, s, top, codes, st); break;
+        case 2: sq8_pf_launch<2>(X, n, d, b, s, top, codes, st); break;
+        case 3: sq8_pf_launch<3>(X, n, d, b, s, top, codes, st); break;
+        case 4: sq8_pf_launch<4>(X, n, d, b, s, top, codes, st); break;
+        case 5: sq8_pf_launch<5>(X, n, d, b, s, top, codes, st); break;
+        case 6: sq8_pf_launch<6>(X, n, d, b, s, top, codes, st); break;
+        case 7: sq8_pf_launch<7>(X, n, d, b, s, top, codes, st); break;
+        default: sq8_pf_launch<8>(X, n, d, b, s, top, codes, st); break;
+        }
+    } else if (v4 && d <= SQ_RS_MAX_D) {
         sq8_encode_rows_kernel<<<grid_for(n * 32, 256), 256, (size_t)d * sizeof(float), st>>>(
             reinterpret_cast<const float4 *>(X), n, d, reinterpret_cast<const float4 *>(b),
             reinterpret_cast<const float4 *>(s), top, reinterpret_cast<uint32_t *>(codes));
@@ -537,10 +624,91 @@ __global__ void rbq1_encode_v4_kernel(const float4 *__restrict__ X, int64_t n, i
     }
 }
 
+// d % 4 == 0 and d <= 1024, NV = ceil(d / 128) float4 per lane, with the next
+// row's loads issued before the current row is evaluated, so every warp always
+// has a row in flight.  Per float4 the four terms of each sum are added plainly
+// and the partial enters the compensated lane sum, so ||r||^2 and ||r||_1 are
+// within about 5 * 2^-24 relative and F within about 12 * 2^-24.
+template <int NV>
+__global__ void __launch_bounds__(256) rbq1_encode_pf_kernel(const float4 *__restrict__ X, int64_t n, int d,
+                                                             const float4 *__restrict__ m,
+                                                             uint32_t *__restrict__ codes, float *__restrict__ nx2,
+                                                             float *__restrict__ F, int32_t *__restrict__ popx) {
+    const int lane = threadIdx.x & 31;
+    const int64_t warp = (blockIdx.x * (int64_t)blockDim.x + threadIdx.x) >> 5;
+    const int64_t nwarps = ((int64_t)gridDim.x * blockDim.x) >> 5;
+    const int W = (d + 31) >> 5, d4 = d >> 2;
+    const float sqrt_d = __fsqrt_rn((float)d);
+    const float4 zero = make_float4(0.0f, 0.0f, 0.0f, 0.0f);
+    float4 cur[NV];
+    auto load_row = [&](int64_t p, float4(&v)[NV]) {
+        const float4 *x = X + p * d4;
+#pragma unroll
+        for (int u = 0; u < NV; ++u) {
+            const int j = 32 * u + lane;
+            v[u] = j < d4 ? __ldg(x + j) : zero;
+        }
+    };
+    if (warp < n) load_row(warp, cur);
+    for (int64_t p = warp; p < n; p += nwarps) {
+        float4 nxt[NV];
+        if (p + nwarps < n) load_row(p + nwarps, nxt);
+        float s2 = 0.0f, c2 = 0.0f, s1 = 0.0f, c1 = 0.0f;
+        int pc = 0;
+#pragma unroll
+        for (int u = 0; u < NV; ++u) {
+            const int j = 32 * u + lane;
+            float4 r = zero;
+            if (j < d4) {
+                const float4 mm = __ldg(m + j);
+                r = make_float4(__fsub_rn(cur[u].x, mm.x), __fsub_rn(cur[u].y, mm.y), __fsub_rn(cur[u].z, mm.z),
+                                __fsub_rn(cur[u].w, mm.w));
+            }
+            // the float4's four terms summed plainly (non-negative terms: relative
+            // error <= 3 * 2^-24), the partial added with compensation
+            kahan_add(s2, c2, __fadd_rn(__fadd_rn(__fmul_rn(r.x, r.x), __fmul_rn(r.y, r.y)),
+                                        __fadd_rn(__fmul_rn(r.z, r.z), __fmul_rn(r.w, r.w))));
+            kahan_add(s1, c1, __fadd_rn(__fadd_rn(fabsf(r.x), fabsf(r.y)), __fadd_rn(fabsf(r.z), fabsf(r.w))));
+            uint32_t nib = (r.x > 0.0f ? 1u : 0u) | (r.y > 0.0f ? 2u : 0u) | (r.z > 0.0f ? 4u : 0u) |
+                           (r.w > 0.0f ? 8u : 0u);
+            nib <<= 4 * (lane & 7);
+            nib |= __shfl_xor_sync(0xffffffffu, nib, 1);
+            nib |= __shfl_xor_sync(0xffffffffu, nib, 2);
+            nib |= __shfl_xor_sync(0xffffffffu, nib, 4);
+            const int wi = 4 * u + (lane >> 3);
+            if ((lane & 7) == 0 && wi < W) {
+                codes[p * W + wi] = nib;
+                pc += __popc(nib);
+            }
+        }
+        rbq1_row_finish(s2, c2, s1, c1, pc, lane, sqrt_d, nx2 + p, F + p, popx + p);
+#pragma unroll
+        for (int u = 0; u < NV; ++u) cur[u] = nxt[u];
+    }
+}
+
+template <int NV>
+static void rbq1_pf_launch(const float *X, int64_t n, int d, const float *m, uint32_t *codes, float *nx2, float *F,
+                           int32_t *popx, cudaStream_t st) {
+    rbq1_encode_pf_kernel<NV><<<grid_for(n * 32, 256), 256, 0, st>>>(
+        reinterpret_cast<const float4 *>(X), n, d, reinterpret_cast<const float4 *>(m), codes, nx2, F, popx);
+}
+
 cudaError_t launch_rbq1_encode(const float *X, int64_t n, int d, const float *m, uint32_t *codes,
                                float *nx2, float *F, int32_t *popx, cudaStream_t st) {
     const int threads = 256;
-    if (d % 4 == 0 && ((uintptr_t)X & 15) == 0 && ((uintptr_t)m & 15) == 0) {
+    if (d % 4 == 0 && d <= 1024 && ((uintptr_t)X & 15) == 0 && ((uintptr_t)m & 15) == 0) {
+        switch ((d + 127) / 128) {
+        case 1: rbq1_pf_launch<1>(X, n, d, m, codes, nx2, F, popx, st); break;
+        case 2: rbq1_pf_launch<2>(X, n, d, m, codes, nx2, F, popx, st); break;
+        case 3: rbq1_pf_launch<3>(X, n, d, m, codes, nx2, F, popx, st); break;
+        case 4: rbq1_pf_launch<4>(X, n, d, m, codes, nx2, F, popx, st); break;
+        case 5: rbq1_pf_launch<5>(X, n, d, m, codes, nx2, F, popx, st); break;
+        case 6: rbq1_pf_launch<6>(X, n, d, m, codes, nx2, F, popx, st); break;
+        case 7: rbq1_pf_launch<7>(X, n, d, m, codes, nx2, F, popx, st); break;
+        default: rbq1_pf_launch<8>(X, n, d, m, codes, nx2, F, popx, st); break;
+        }
+    } else if (d % 4 == 0 && ((uintptr_t)X & 15) == 0 && ((uintptr_t)m & 15) == 0) {
         rbq1_encode_v4_kernel<<<grid_for(n * 32, threads), threads, 0, st>>>(
             reinterpret_cast<const float4 *>(X), n, d, reinterpret_cast<const float4 *>(m), codes, nx2, F,
             popx);

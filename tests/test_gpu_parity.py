@@ -280,7 +280,8 @@ def _rbq1_host(r):
     return h
 
 
-@pytest.mark.parametrize("n,d", [(3000, 768), (777, 33), (500, 32), (400, 31), (100, 1), (333, 36), (257, 1500)])
+@pytest.mark.parametrize("n,d", [(3000, 768), (777, 33), (500, 32), (400, 31), (100, 1), (333, 36), (257, 1500),
+                                 (5000, 1024), (4999, 516)])
 def test_encode_rbq1_vs_oracle(skm, n, d):
     X = _points(n, d, seed=n + 1)
     r = skm.skm_quantize(skm.REPR_RBQ1, X.to(DEV))
