@@ -62,6 +62,14 @@ enum { MODE_SCREEN = 0, MODE_SQ8 = 1, MODE_RBQ1 = 2, MODE_LVQ4 = 3, MODE_GEMM = 
 // at 1M x 1000 x 768), so every mode runs one CTA per cluster.
 constexpr int TC_NH[5] = {4, 2, 4, 4, 4};
 constexpr int TC_CL[5] = {1, 1, 1, 1, 1};
+// Job streams per CTA, by mode.  NS = 2: the CTA's point tiles form two
+// streams whose jobs the MMA warp issues alternately, each into its own TMEM
+// accumulator, each drained by its own half of the epilogue warps; an
+// epilogue group then has two MMA jobs' time per job.  NS = 1: one stream, the
+// two accumulators alternate by job and every epilogue warp takes every job.
+// (NS = 2 needs at least 256 epilogue threads per group for the e4m3 and SQ8
+// records.)
+constexpr int TC_NS[5] = {2, 1, 2, 2, 2};
 // GEMM mode (the projection Y = (X - mean) P in fp32 accuracy from bf16
 // parts x = x1 + x2 + x3, P = p1 + p2 + p3): K segments of (A part, B part),
 // the smallest products first; parts i + j > 4 (below 2^-24 relative) are left
@@ -93,11 +101,12 @@ constexpr int merge_words() { return MODE == MODE_SCREEN ? 2 * TCAND + 2 : 2; }
 // double-buffered by job.
 constexpr int REC_BYTES = 4096;
 // 1024-byte alignment slack, the stages, barriers + TMEM slot (352 bytes), the
-// merge buffer (slices 1..NH-1 publish) and the record buffers.
-template <int MODE, int NH>
+// merge buffer (per group, slices 1..NH/NS-1 publish) and the record buffers
+// (two per group).
+template <int MODE, int NH, int NS>
 constexpr size_t tc_smem_bytes() {
     return 1024 + (size_t)STAGES * (A_STAGE + B_STAGE) + 512 +
-           (size_t)(NH - 1) * BM * merge_words<MODE>() * 4 + 2 * REC_BYTES;
+           (size_t)(NH - NS) * BM * merge_words<MODE>() * 4 + 2 * NS * REC_BYTES;
 }
 
 struct TcParams {
@@ -438,10 +447,13 @@ __device__ __forceinline__ void ct_range(const TcParams &p, int64_t rt, int &lo,
     }
 }
 
-template <int MODE, int NH, int CL, bool SEG>
+template <int MODE, int NH, int CL, bool SEG, int NS>
 __global__ void __launch_bounds__(tc_threads<NH>(), 1)
     tc_assign_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                      const TcParams p) {
+    static_assert(NS == 1 || (NS == 2 && CL == 1 && NH % 2 == 0), "two job streams: one CTA per cluster");
+    static_assert(NS == 1 || MODE == MODE_GEMM || epi_threads<NH>() / NS >= (MODE == MODE_SCREEN ? 128 : 256),
+                  "records staged by one epilogue group");
     extern __shared__ uint8_t smem_raw[];
     const uint32_t raw = smem_u32(smem_raw);
     const uint32_t base = (raw + 1023u) & ~1023u;
@@ -469,7 +481,7 @@ __global__ void __launch_bounds__(tc_threads<NH>(), 1)
         }
         for (int b = 0; b < 2; ++b) {
             mbar_init(tfull_bar(b), 1);
-            mbar_init(tempty_bar(b), epi_threads<NH>());
+            mbar_init(tempty_bar(b), epi_threads<NH>() / NS);
         }
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
         asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmA)) : "memory");
@@ -499,14 +511,68 @@ __global__ void __launch_bounds__(tc_threads<NH>(), 1)
     const int64_t ngroups = (p.nrt + CL - 1) / CL;
     if (CL > 1) cluster_sync_all();  // peers' barriers are initialised before any multicast
 
+    // Job order (producer and MMA issuer walk it identically): stream s takes
+    // the CTA's point-tile groups g0 + (s + NS i) gstep; the streams' jobs
+    // (point tile, centroid tile) are issued round-robin.
+    struct JobStream {
+        int64_t g;
+        int ct, hi;
+    };
+    auto stream_seek = [&](JobStream &js) {  // the first job at or after group js.g
+        while (js.g < ngroups) {
+            int lo, hi;
+            ct_range(p, js.g * CL + crank, lo, hi);
+            if (lo < hi) {
+                js.ct = lo;
+                js.hi = hi;
+                return;
+            }
+            js.g += NS * gstep;
+        }
+    };
+    auto stream_advance = [&](JobStream &js) {
+        if (++js.ct >= js.hi) {
+            js.g += NS * gstep;
+            stream_seek(js);
+        }
+    };
+    // the stream of the next job (turn first), or -1 when both are done;
+    // streams are indexed by constants only, so they stay in registers
+    auto stream_g = [&](const JobStream(&js)[NS], int s) { return s == 0 ? js[0].g : js[NS - 1].g; };
+    auto stream_pick = [&](const JobStream(&js)[NS], int turn) {
+        if (stream_g(js, turn) < ngroups) return turn;
+        const int o = (turn + 1) % NS;
+        return stream_g(js, o) < ngroups ? o : -1;
+    };
+    auto stream_take = [&](JobStream(&js)[NS], int s, int64_t &g, int &ct) {  // the job, then advance
+        if (s == 0) {
+            g = js[0].g;
+            ct = js[0].ct;
+            stream_advance(js[0]);
+        } else {
+            g = js[NS - 1].g;
+            ct = js[NS - 1].ct;
+            stream_advance(js[NS - 1]);
+        }
+    };
+
     if (warp == 0) {
         if (lane == 0) {  // ---------------------------------------- TMA producer
             uint32_t it = 0;
-            for (int64_t g = g0; g < ngroups; g += gstep) {
-                const int64_t rt = g * CL + crank;
-                int ct_lo, ct_hi;
-                ct_range(p, rt, ct_lo, ct_hi);
-                for (int ct = ct_lo; ct < ct_hi; ++ct)
+            JobStream js[NS];
+            for (int s = 0; s < NS; ++s) {
+                js[s].g = g0 + s * gstep;
+                stream_seek(js[s]);
+            }
+            for (int turn = 0;;) {
+                const int sj = stream_pick(js, turn);
+                if (sj < 0) break;
+                int64_t gj;
+                int ct;
+                stream_take(js, sj, gj, ct);
+                const int64_t rt = gj * CL + crank;
+                turn = (sj + 1) % NS;
+                {
                     for (int kt = 0; kt < NSEG * p.nkc; ++kt, ++it) {
                         const int seg = kt / p.nkc, kc = kt - seg * p.nkc;
                         const int arow = (int)(rt * BM) + (NSEG > 1 ? GEMM_SEG_A[seg] * (int)p.n : 0);
@@ -522,17 +588,34 @@ __global__ void __launch_bounds__(tc_threads<NH>(), 1)
                                            ct * BN + (int)crank * (BN / CL), full_bar(s),
                                            (uint16_t)((1u << CL) - 1u));
                     }
+                }
             }
         producer_done:;
         }
     } else if (warp == 1) {
         if (lane == 0) {  // ---------------------------------------- MMA issuer
             uint32_t it = 0, job = 0;
-            for (int64_t g = g0; g < ngroups; g += gstep) {
-                int ct_lo, ct_hi;
-                ct_range(p, g * CL + crank, ct_lo, ct_hi);
-                for (int ct = ct_lo; ct < ct_hi; ++ct, ++job) {
-                    const uint32_t b = job & 1u, bph = (job >> 1) & 1u;
+            uint32_t jc[NS];
+            JobStream js[NS];
+            for (int s = 0; s < NS; ++s) {
+                js[s].g = g0 + s * gstep;
+                jc[s] = 0;
+                stream_seek(js[s]);
+            }
+            for (int turn = 0;; ++job) {
+                const int sj = stream_pick(js, turn);
+                if (sj < 0) break;
+                {
+                    int64_t gj;
+                    int ctj;
+                    stream_take(js, sj, gj, ctj);
+                }
+                turn = (sj + 1) % NS;
+                {
+                    // NS = 2: stream sj owns accumulator sj; NS = 1: they alternate
+                    const uint32_t b = NS == 2 ? (uint32_t)sj : (job & 1u);
+                    const uint32_t use = sj == 0 ? jc[0]++ : jc[NS - 1]++;
+                    const uint32_t bph = NS == 2 ? (use & 1u) : ((job >> 1) & 1u);
                     if (!mbar_wait(tempty_bar(b), bph ^ 1u, abort_flag)) goto mma_done;
                     tc_fence_after();
                     const uint32_t dcol = tmem + b * BN;
@@ -560,21 +643,27 @@ __global__ void __launch_bounds__(tc_threads<NH>(), 1)
         mma_done:;
         }
     } else {  // ------------------------------------------------------- epilogue
-        constexpr int SW = BN / NH;      // columns per slice
+        constexpr int NHG = NH / NS;     // warps per TMEM lane quarter in a group
+        constexpr int GT = epi_threads<NH>() / NS;  // threads per group
+        constexpr int SW = BN / NHG;     // columns per slice
         constexpr int MW = merge_words<MODE>();
         const int e = warp - 2;          // 0 .. 4 NH - 1
         const int q = warp & 3;          // TMEM lane quarter this warp may access
-        const int slice = e >> 2;        // which SW of the 256 columns
+        const int grp = (e >> 2) / NHG;  // job stream (and accumulator) of this warp
+        const int slice = (e >> 2) % NHG;  // which SW of the 256 columns
         const int rin = q * 32 + lane;   // row within the point tile
-        uint32_t *merge = reinterpret_cast<uint32_t *>(tmem_slot + 64);  // [NH-1][BM][MW]
+        // per group [NHG-1][BM][MW]
+        uint32_t *merge = reinterpret_cast<uint32_t *>(tmem_slot + 64) + (size_t)grp * (NHG - 1) * BM * MW;
         // Records of the job's 256 centroids (SCREEN: 128 ||c||^2 pairs; RBQ1:
         // 128 rinfo + 128 rinfoq pairs; SQ8: 256 nc), copied into
         // shared memory at the start of each job from registers that were
         // loaded one job ahead, so the per-column reads are shared-memory
         // broadcasts.  Buffer (job & 1) is rewritten only after every epilogue
         // thread has passed the next job's barrier, i.e. finished reading it.
-        uint8_t *rec_base = reinterpret_cast<uint8_t *>(merge + (NH - 1) * BM * MW);
-        const int te = threadIdx.x - 64;  // 0 .. epi_threads - 1
+        uint8_t *rec_base = reinterpret_cast<uint8_t *>(reinterpret_cast<uint32_t *>(tmem_slot + 64) +
+                                                        (size_t)(NH - NS) * BM * MW) +
+                            (size_t)grp * 2 * REC_BYTES;  // this group's two buffers
+        const int te = threadIdx.x - 64 - grp * GT;  // 0 .. GT - 1
         float4 pre4 = make_float4(0.f, 0.f, 0.f, 0.f);
         float2 pre2 = make_float2(0.f, 0.f);
         int32_t pre1 = 0;
@@ -603,14 +692,14 @@ __global__ void __launch_bounds__(tc_threads<NH>(), 1)
         };
         {
             int lo0, hi0;
-            ct_range(p, g0 * CL + crank, lo0, hi0);
+            ct_range(p, (g0 + grp * gstep) * CL + crank, lo0, hi0);
             rec_load(lo0);
         }
         // A warp whose barrier wait gave up stops computing but keeps taking part
         // in the named barriers, so the other epilogue warps never wait on it.
         bool dead = false;
-        uint32_t job = 0;
-        for (int64_t g = g0; g < ngroups; g += gstep) {
+        uint32_t job = 0;  // jobs of this group so far (NS = 1: of the CTA)
+        for (int64_t g = g0 + grp * gstep; g < ngroups; g += NS * gstep) {
             const int64_t rt = g * CL + crank;
             const int64_t row = rt * BM + rin;
             const bool valid = row < p.n;
@@ -633,7 +722,7 @@ __global__ void __launch_bounds__(tc_threads<NH>(), 1)
             int next_lo = 0;
             {
                 int nhi;
-                ct_range(p, (g + gstep) * CL + crank, next_lo, nhi);
+                ct_range(p, (g + NS * gstep) * CL + crank, next_lo, nhi);
             }
             if (MODE == MODE_SCREEN) {
                 a2 = valid ? 2.0f * p.xinfo[row].x : 0.0f;
@@ -654,16 +743,20 @@ __global__ void __launch_bounds__(tc_threads<NH>(), 1)
                 rpc = valid ? (float)(2 * p.popx[row] - p.d) : 0.0f;
             }
             for (int ct = ct_lo; ct < ct_hi; ++ct, ++job) {
-                const uint32_t b = job & 1u, bph = (job >> 1) & 1u;
+                // accumulator b (NS = 2: the group's own; NS = 1: alternating), its
+                // use parity, and the record buffer (two per group, alternating)
+                const uint32_t b = NS == 2 ? (uint32_t)grp : (job & 1u);
+                const uint32_t bph = NS == 2 ? (job & 1u) : ((job >> 1) & 1u);
+                const uint32_t rb = job & 1u;
                 bool ok = true;
                 if (!dead) ok = mbar_wait(tfull_bar(b), bph, abort_flag);
                 dead = dead || !__all_sync(0xffffffffu, ok);
-                rec_store(b);
-                asm volatile("bar.sync 2, %0;" ::"n"(epi_threads<NH>()) : "memory");
+                rec_store(rb);
+                asm volatile("bar.sync %0, %1;" ::"r"(2 + grp), "n"(GT) : "memory");
                 rec_load(ct + 1 < ct_hi ? ct + 1 : next_lo);
                 if (dead) continue;
                 tc_fence_after();
-                const uint8_t *rbuf = rec_base + b * REC_BYTES;
+                const uint8_t *rbuf = rec_base + rb * REC_BYTES;
                 const uint32_t taddr = tmem + ((uint32_t)(q * 32) << 16) + b * BN + slice * SW;
                 const int jh = ct * BN + slice * SW;
                 if (MODE == MODE_GEMM) {
@@ -928,11 +1021,11 @@ __global__ void __launch_bounds__(tc_threads<NH>(), 1)
                     slot[1] = (uint32_t)besti;
                 }
             }
-            asm volatile("bar.sync 1, %0;" ::"n"(epi_threads<NH>()) : "memory");
+            asm volatile("bar.sync %0, %1;" ::"r"(NS == 2 ? 4 + grp : 1), "n"(GT) : "memory");
             if (slice == 0 && valid && !dead) {
                 // slices in increasing column order; ties resolve to the lower index
 #pragma unroll
-                for (int h = 1; h < NH; ++h) {
+                for (int h = 1; h < NHG; ++h) {
                     const uint32_t *slot = merge + ((h - 1) * BM + rin) * MW;
                     if (MODE == MODE_SCREEN) {
                         sr.umin = fminf(sr.umin, __uint_as_float(slot[2 * TCAND]));
@@ -1452,9 +1545,10 @@ int launch_tc(const void *xs, int64_t n, int dp, int d, const void *cs, int k, c
               cudaStream_t st) {
     constexpr int NH = TC_NH[MODE];
     constexpr int CL = TC_CL[MODE];
-    constexpr size_t SMEM = tc_smem_bytes<MODE, NH>();
+    constexpr int NS = TC_NS[MODE];
+    constexpr size_t SMEM = tc_smem_bytes<MODE, NH, NS>();
     static_assert(SMEM <= 227 * 1024, "shared memory per CTA");
-    auto kern = p0.seg_group ? tc_assign_kernel<MODE, NH, CL, true> : tc_assign_kernel<MODE, NH, CL, false>;
+    auto kern = p0.seg_group ? tc_assign_kernel<MODE, NH, CL, true, NS> : tc_assign_kernel<MODE, NH, CL, false, NS>;
     const int segi = p0.seg_group ? 1 : 0;
     // per device: the attribute and the number of clusters that fit at once
     constexpr int MAXDEV = 64;
