@@ -451,10 +451,18 @@ def run_ours(args):
             t = torch.tensor([ems], device=dev, dtype=torch.float64)
             dist.all_reduce(t, op=dist.ReduceOp.MAX)
             ems = float(t.item())
+        # and right after it: the link is shared with the host's other traffic
+        torch.cuda.synchronize()
+        p0.record(stream)
+        Xbuf[0].copy_(X_host, non_blocking=True)
+        p1.record(stream)
+        torch.cuda.synchronize()
+        h2d_probe_after_gbs = X_host.numel() * 4 / (p0.elapsed_time(p1) / 1e3) / 1e9
         e2e = {"value": world * 2.0 * N_POINTS * K * e2e_steps / (ems / 1e3), "unit": "distances/s",
                "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "steps": e2e_steps,
                "host_enqueue_ms_per_step": round(statistics.mean(host_ms), 3),
-               "h2d_probe_gbs": round(h2d_probe_gbs, 1),
+               "h2d_probe_gbs": round(h2d_probe_gbs, 1), "h2d_probe_after_gbs": round(h2d_probe_after_gbs, 1),
+               "h2d_effective_gbs": round(h2d / (ems / e2e_steps / 1e3) / 1e9, 1),
                "ms_per_step": ems / e2e_steps,
                "path": f"pinned host fp32 points -> H2D in {nchunk} row ranges on a copy stream (two device "
                        "buffers: the next step's points stream in during this step's tail), each range assigned "

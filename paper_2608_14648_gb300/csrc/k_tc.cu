@@ -60,7 +60,7 @@ enum { MODE_SCREEN = 0, MODE_SQ8 = 1, MODE_RBQ1 = 2, MODE_LVQ4 = 3, MODE_GEMM = 
 // correctly but measured slower on GB300 (the pair's pipelines wait on each
 // other's slowest epilogue: fp32 0.999 vs 0.956 ms, 1-bit 0.602 vs 0.554 ms
 // at 1M x 1000 x 768), so every mode runs one CTA per cluster.
-constexpr int TC_NH[5] = {4, 2, 4, 4, 4};
+constexpr int TC_NH[5] = {4, 4, 4, 4, 4};
 constexpr int TC_CL[5] = {1, 1, 1, 1, 1};
 // Job streams per CTA, by mode.  NS = 2: the CTA's point tiles form two
 // streams whose jobs the MMA warp issues alternately, each into its own TMEM
@@ -68,8 +68,10 @@ constexpr int TC_CL[5] = {1, 1, 1, 1, 1};
 // epilogue group then has two MMA jobs' time per job.  NS = 1: one stream, the
 // two accumulators alternate by job and every epilogue warp takes every job.
 // (NS = 2 needs at least 256 epilogue threads per group for the e4m3 and SQ8
-// records.)
-constexpr int TC_NS[5] = {2, 1, 2, 2, 2};
+// records.)  Measured at 1M x 1000 x 768 against one stream: 1-bit 0.508 vs
+// 0.574 ms, LVQ4 0.532 vs 0.575, fp32 screen 0.99 vs 1.02, SQ8 (with NH = 4)
+// 0.847 vs 0.882.
+constexpr int TC_NS[5] = {2, 2, 2, 2, 2};
 // GEMM mode (the projection Y = (X - mean) P in fp32 accuracy from bf16
 // parts x = x1 + x2 + x3, P = p1 + p2 + p3): K segments of (A part, B part),
 // the smallest products first; parts i + j > 4 (below 2^-24 relative) are left
@@ -79,8 +81,10 @@ __device__ constexpr int GEMM_SEG_A[GEMM_NSEG] = {2, 1, 0, 1, 0, 0};
 __device__ constexpr int GEMM_SEG_B[GEMM_NSEG] = {0, 1, 2, 0, 1, 0};
 // Columns per TMEM load in the e4m3 epilogues (32: one load and wait per 32
 // columns; 16: two buffers, the next load in flight).  Measured on GB300 at
-// 1M x 1000 x 768: 16 is 1-3% faster for both e4m3 modes.
-constexpr int F8_CW = 16;
+// 1M x 1000 x 768 with two job streams: 16 for the 1-bit epilogue (0.511 vs
+// 0.529 ms), 32 for LVQ4 (0.516 vs 0.531 ms).
+template <int MODE>
+constexpr int f8_cw() { return MODE == 3 /* MODE_LVQ4 */ ? 32 : 16; }
 // The same choice for the fp32 / bf16 screen's epilogue, whose pass 1 is one
 // packed FMA per column pair: 32 is 2-4% faster there (C1 1.014 vs 1.032 ms,
 // C4 38.1 vs 39.7 ms).
@@ -892,6 +896,7 @@ __global__ void __launch_bounds__(tc_threads<NH>(), 1)
                 } else if (f8_mode<MODE>()) {
                     // e4m3 modes: chunks of F8_CW columns (F8_CW = 16: the next
                     // chunk's TMEM load in flight while this one is evaluated)
+                    constexpr int F8_CW = f8_cw<MODE>();
                     constexpr int NC = SW / F8_CW;
                     constexpr int G = F8_CW / 8;
                     auto chunk = [&](const uint32_t(&v)[F8_CW], int c) {
