@@ -1,18 +1,19 @@
 // Tensor-core assignment (Section 2.3 STEP 2 "GEMM of the data points and
 // centroids", Section 3.1 8-bit GEMM) on sm_103a with tcgen05 + TMEM + TMA.
 //
-// One persistent CTA per SM walks (point tile, centroid tile) jobs:
+// One persistent CTA per SM walks (point tile, centroid tile) jobs; its point
+// tiles form two job streams whose jobs are issued alternately:
 //   warp 0      TMA producer: 128 x 64 point slice and 256 x 64 centroid slice
 //               (bf16, 128-byte swizzle) per stage, 4-stage mbarrier ring
 //   warp 1      MMA issuer: 4 x tcgen05.mma.kind::f16 (M=128, N=256, K=16)
-//               per stage into one of two 128 x 256 fp32 TMEM accumulators
-//   warps 2..   epilogue: tcgen05.ld of the accumulator (thread = point row;
-//               NH warps per TMEM lane quarter, each taking 256 / NH of the
-//               columns), fused per-row reduction over centroids, so the
-//               N x K distance matrix never leaves the SM; the NH column
-//               slices of a row merge through shared memory at the end of a
-//               point tile
-// Two epilogues:
+//               per stage into the stream's 128 x 256 fp32 TMEM accumulator
+//   warps 2..   epilogue, one group of warps per stream: tcgen05.ld of the
+//               accumulator (thread = point row; NH / 2 warps per TMEM lane
+//               quarter, each taking a slice of the columns), fused per-row
+//               reduction over centroids, so the N x K distance matrix never
+//               leaves the SM; the column slices of a row merge through
+//               shared memory at the end of its point tile
+// Epilogues:
 //  SCREEN (fp32 / bf16 points): bf16 operands, so the dot product carries a
 //    rounding error.  Each pair gets a rigorous interval [L, U] for
 //    s = ||c||^2 - 2 x.c (the distance minus ||x||^2) from per-row and
