@@ -42,8 +42,8 @@ POPC_PER_CLK_SM = 16
 # capture each (200,000 points x d=768, k=1000; profiles/tc_assign_*.md).
 # Each point row is read once per launch, so traffic scales with the points.
 TRAFFIC_PER_POINT = {
-    "assign_f32": (311.921408e6 + 5.200896e6) / 200_000,
-    "assign_rbq1": (156.846848e6 + 3.305728e6) / 200_000,
+    "assign_f32": (314.849280e6 + 5.701888e6) / 200_000,
+    "assign_rbq1": (156.890624e6 + 3.590912e6) / 200_000,
 }
 
 
