@@ -428,11 +428,22 @@ def run_ours(args):
                     skm.skm_quantize(skm.REPR_RBQ1, xb[b0:b1], fit=False, m=mE, ws=wsQ2, out=qo)
                     skm.skm_assign(prc, CdR, K, want_dist=False, ws=wsAR2, out=aR[b0:b1])
                 buf_free[slot].record(stream)
+                if world > 1:  # the same exchange as the device-resident step
+                    skd.allreduce_partials(part32e, cnt32e)
                 skm.skm_update_finalize(pall[slot], part32e, cnt32e, Cd32)
                 host_ms.append((time.perf_counter() - th0) * 1e3)  # enqueue only (no sync so far)
                 eE = skm.skm_rbq1_exponent(FE)
+                if world > 1:
+                    eE = skd.global_exponent(eE, dev)
                 pR2 = skm.Points(skm.REPR_RBQ1, codesE, DIM, nx2E, FE, popxE, mE, eE)
-                skm.skm_update(pR2, aR, CdR, counts=cntR, ws=wsUR)
+                if world > 1:
+                    partR.zero_()
+                    cntR.zero_()
+                    skm.skm_update(pR2, aR, None, counts=cntR, partial=partR, ws=wsUR)
+                    skd.allreduce_partials(partR, cntR)
+                    skm.skm_update_finalize(pR2, partR, cntR, CdR)
+                else:
+                    skm.skm_update(pR2, aR, CdR, counts=cntR, ws=wsUR)
                 a_host[0].copy_(a32, non_blocking=True)
                 a_host[1].copy_(aR, non_blocking=True)
                 C_host32.copy_(Cd32, non_blocking=True)

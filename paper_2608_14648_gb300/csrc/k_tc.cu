@@ -60,7 +60,9 @@ enum { MODE_SCREEN = 0, MODE_SQ8 = 1, MODE_RBQ1 = 2, MODE_LVQ4 = 3, MODE_GEMM = 
 // slices multicast across the cluster), by mode.  Clusters of 2 run
 // correctly but measured slower on GB300 (the pair's pipelines wait on each
 // other's slowest epilogue: fp32 0.999 vs 0.956 ms, 1-bit 0.602 vs 0.554 ms
-// at 1M x 1000 x 768), so every mode runs one CTA per cluster.
+// at 1M x 1000 x 768 with one job stream; with two job streams 1-bit 0.516
+// vs 0.512 ms, LVQ4 0.537 vs 0.516 ms), so every mode runs one CTA per
+// cluster.  Segmented mode always does.
 constexpr int TC_NH[5] = {4, 4, 4, 4, 4};
 constexpr int TC_CL[5] = {1, 1, 1, 1, 1};
 // Job streams per CTA, by mode.  NS = 2: the CTA's point tiles form two
@@ -456,7 +458,8 @@ template <int MODE, int NH, int CL, bool SEG, int NS>
 __global__ void __launch_bounds__(tc_threads<NH>(), 1)
     tc_assign_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                      const TcParams p) {
-    static_assert(NS == 1 || (NS == 2 && CL == 1 && NH % 2 == 0), "two job streams: one CTA per cluster");
+    static_assert(NS == 1 || (NS == 2 && NH % 2 == 0), "two job streams: two epilogue groups");
+    static_assert(CL == 1 || !SEG, "segmented mode: one CTA per cluster");
     static_assert(NS == 1 || MODE == MODE_GEMM || epi_threads<NH>() / NS >= (MODE == MODE_SCREEN ? 128 : 256),
                   "records staged by one epilogue group");
     extern __shared__ uint8_t smem_raw[];
@@ -1546,16 +1549,28 @@ int device_sms() {
     return sms > 0 ? sms : 148;
 }
 
+// Segmented mode runs one CTA per cluster: the CTAs of a cluster would walk
+// different centroid ranges, so there is no common slice to multicast.
+template <int MODE, int CL, bool SEG>
+int launch_tc_cl(const void *xs, int64_t n, int dp, int d, const void *cs, int k, const TcParams &p0,
+                 cudaStream_t st);
+
 template <int MODE>
 int launch_tc(const void *xs, int64_t n, int dp, int d, const void *cs, int k, const TcParams &p0,
               cudaStream_t st) {
+    if (p0.seg_group) return launch_tc_cl<MODE, 1, true>(xs, n, dp, d, cs, k, p0, st);
+    return launch_tc_cl<MODE, TC_CL[MODE], false>(xs, n, dp, d, cs, k, p0, st);
+}
+
+template <int MODE, int CL, bool SEG>
+int launch_tc_cl(const void *xs, int64_t n, int dp, int d, const void *cs, int k, const TcParams &p0,
+                 cudaStream_t st) {
     constexpr int NH = TC_NH[MODE];
-    constexpr int CL = TC_CL[MODE];
     constexpr int NS = TC_NS[MODE];
     constexpr size_t SMEM = tc_smem_bytes<MODE, NH, NS>();
     static_assert(SMEM <= 227 * 1024, "shared memory per CTA");
-    auto kern = p0.seg_group ? tc_assign_kernel<MODE, NH, CL, true, NS> : tc_assign_kernel<MODE, NH, CL, false, NS>;
-    const int segi = p0.seg_group ? 1 : 0;
+    auto kern = tc_assign_kernel<MODE, NH, CL, SEG, NS>;
+    const int segi = SEG ? 1 : 0;
     // per device: the attribute and the number of clusters that fit at once
     constexpr int MAXDEV = 64;
     static std::mutex mu;
