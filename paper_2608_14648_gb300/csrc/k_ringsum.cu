@@ -441,6 +441,15 @@ struct Sq8Cons {
         cur = __shfl_sync(0xffffffffu, clw, 0);
     }
     __device__ __forceinline__ void row(int i, const uint8_t *slot, int lane) {
+        uint4 w[NG];
+        const int ng16 = d >> 4;  // 16-byte groups (d % 16 == 0 on this path)
+#pragma unroll
+        for (int t = 0; t < NG; ++t)
+            if (lane + 32 * t < ng16) w[t] = reinterpret_cast<const uint4 *>(slot)[lane + 32 * t];
+        row_regs(i, w, lane);
+    }
+    // the same with the lane's 16-byte groups of the row already in registers
+    __device__ __forceinline__ void row_regs(int i, const uint4 (&wr)[NG], int lane) {
         if ((i & 31) == 0 && i > 0) {
             clw = cln;
             const int nx = i + 32 + lane;
@@ -451,12 +460,12 @@ struct Sq8Cons {
             flush(cur, lane);
             cur = c;
         }
-        const int ng16 = d >> 4;  // 16-byte groups (d % 16 == 0 on this path)
+        const int ng16 = d >> 4;
 #pragma unroll
         for (int t = 0; t < NG; ++t) {
             const int gidx = lane + 32 * t;
             if (gidx < ng16) {
-                const uint4 w = reinterpret_cast<const uint4 *>(slot)[gidx];
+                const uint4 w = wr[t];
                 ev[4 * t + 0] += w.x & 0x00ff00ffu;
                 od[4 * t + 0] += (w.x >> 8) & 0x00ff00ffu;
                 ev[4 * t + 1] += w.y & 0x00ff00ffu;
@@ -483,6 +492,55 @@ __global__ void __launch_bounds__(RS_THREADS) ring_sum_sq8_kernel(
     cons.S = S;
     cons.d = d;
     ring_gather(codes, perm, nval, L, flag, cons);
+}
+
+// SQ8 rows of at most 1 KB, read straight into registers: no ring.  Lane l
+// loads the 16-byte groups l + 32 t of a row with 128-bit loads; the loads of
+// the next SQ8_PF rows of the warp's run are in flight while a row is summed
+// (a row's slot in the register buffer is refilled right after it is read),
+// and with little shared memory many warps fit per SM.
+constexpr int SQ8_PF = 4;
+template <int NG>
+__global__ void __launch_bounds__(RS_THREADS) direct_sum_sq8_kernel(
+    const uint8_t *__restrict__ codes, int d, const int32_t *__restrict__ perm,
+    const int32_t *__restrict__ scl, const int64_t *__restrict__ offsets, int k,
+    unsigned long long *__restrict__ S) {
+    __shared__ int32_t sperm_all[RS_CW][RS_ROWS];
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int64_t nval = offsets[k];
+    const int64_t q0 = ((int64_t)blockIdx.x * RS_CW + warp) * RS_ROWS;
+    const int cnt = run_len(nval, q0);
+    if (cnt == 0) return;
+    int32_t *sperm = sperm_all[warp];
+    for (int i = lane; i < cnt; i += 32) sperm[i] = perm[q0 + i];
+    __syncwarp();
+    const int ng16 = d >> 4;
+    auto load = [&](int r, uint4(&w)[NG]) {
+        const uint4 *src = reinterpret_cast<const uint4 *>(codes + (size_t)sperm[r] * d);
+#pragma unroll
+        for (int t = 0; t < NG; ++t)
+            if (lane + 32 * t < ng16) w[t] = __ldg(src + lane + 32 * t);
+    };
+    Sq8Cons<NG> cons;
+    cons.scl = scl;
+    cons.S = S;
+    cons.d = d;
+    uint4 buf[SQ8_PF][NG];
+#pragma unroll
+    for (int p = 0; p < SQ8_PF; ++p)
+        if (p < cnt) load(p, buf[p]);
+    cons.start(q0, cnt, lane);
+    for (int r0 = 0; r0 < cnt; r0 += SQ8_PF) {
+#pragma unroll
+        for (int p = 0; p < SQ8_PF; ++p) {
+            const int r = r0 + p;
+            if (r < cnt) {  // warp-uniform
+                cons.row_regs(r, buf[p], lane);
+                if (r + SQ8_PF < cnt) load(r + SQ8_PF, buf[p]);
+            }
+        }
+    }
+    cons.finish(lane);
 }
 
 // ------------------------------------------------------------- LVQ4 rows
@@ -739,6 +797,13 @@ cudaError_t launch_ring_sum_sq8(const uint8_t *codes, int64_t n, int d, const in
     const unsigned g = ring_blocks(n);
     auto S64 = reinterpret_cast<unsigned long long *>(S);
     const int q = (d / 16 + 31) / 32;  // 16-byte groups per lane
+    if (d <= 1024) {  // rows of at most 1 KB: straight into registers
+        if (q <= 1)
+            direct_sum_sq8_kernel<1><<<g, RS_THREADS, 0, st>>>(codes, d, perm, scl, offsets, k, S64);
+        else
+            direct_sum_sq8_kernel<2><<<g, RS_THREADS, 0, st>>>(codes, d, perm, scl, offsets, k, S64);
+        return launched();
+    }
 #define RS_CASE(NGV)                                                                                \
     if (q <= NGV) {                                                                                 \
         auto kern = ring_sum_sq8_kernel<NGV>;                                                       \
