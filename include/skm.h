@@ -41,7 +41,7 @@ extern "C" {
 typedef enum skm_status {
     SKM_OK = 0,
     SKM_ERR_INVALID_ARG = 1,  /* bad shape, null pointer, k > n, bad enum    */
-    SKM_ERR_UNSUPPORTED = 2,  /* valid but outside this build's limits       */
+    SKM_ERR_UNSUPPORTED = 2,  /* valid but outside the library's limits     */
     SKM_ERR_CUDA = 3,         /* a CUDA runtime/driver call failed            */
     SKM_ERR_NO_MEMORY = 4,    /* ws_bytes smaller than skm_workspace_size()  */
     SKM_ERR_TIMEOUT = 5,      /* a bounded device wait gave up               */
