@@ -44,36 +44,47 @@ cudaError_t launch_histogram(const int32_t *assign, int64_t n, int k, int32_t *c
     if (n == 0) return cudaSuccess;
     const int use_smem = k <= 12288;
     const size_t smem = use_smem ? sizeof(int32_t) * (size_t)k : 0;
-    int64_t blocks = (n + 1023) / 1024;
-    if (blocks > 152 * 4) blocks = 152 * 4;
-    histogram_kernel<<<(unsigned)blocks, 512, smem, st>>>(assign, n, k, counts32, use_smem);
+    // few blocks: each one adds its nonzero shared counters to the global ones,
+    // so the global atomics grow with blocks x k
+    int64_t blocks = (n + 4095) / 4096;
+    if (blocks > 152 * 2) blocks = 152 * 2;
+    histogram_kernel<<<(unsigned)blocks, 1024, smem, st>>>(assign, n, k, counts32, use_smem);
     return launched();
 }
 
 // --------------------------------------------------------------------- scan
-// Single block; each thread scans a contiguous run of counts.
+// Single block of 1024 threads; each thread scans a contiguous run of counts.
 __global__ void scan_offsets_kernel(const int32_t *__restrict__ counts, int k,
                                     int64_t *__restrict__ offsets, int64_t *__restrict__ counts64,
                                     int accumulate) {
-    __shared__ int64_t part[1024];
-    const int t = threadIdx.x;
+    __shared__ int64_t wsum[32];
+    const int t = threadIdx.x, lane = t & 31, w = t >> 5;
     const int per = (k + blockDim.x - 1) / blockDim.x;
     const int lo = min(k, t * per), hi = min(k, lo + per);
     int64_t s = 0;
     for (int j = lo; j < hi; ++j) s += counts[j];
-    part[t] = s;
+    // exclusive scan of the threads' run sums: shuffles inside each warp, then
+    // the warp totals (exact integer sums, so any order gives the same offsets)
+    int64_t v = s;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+        const int64_t u = __shfl_up_sync(0xffffffffu, v, o);
+        if (lane >= o) v += u;
+    }
+    if (lane == 31) wsum[w] = v;
     __syncthreads();
-    if (t == 0) {
-        int64_t run = 0;
-        for (int i = 0; i < (int)blockDim.x; ++i) {
-            const int64_t v = part[i];
-            part[i] = run;
-            run += v;
+    if (w == 0) {
+        int64_t x = lane < (int)(blockDim.x >> 5) ? wsum[lane] : 0;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+            const int64_t u = __shfl_up_sync(0xffffffffu, x, o);
+            if (lane >= o) x += u;
         }
-        offsets[k] = run;
+        wsum[lane] = x;  // inclusive over warps
     }
     __syncthreads();
-    int64_t run = part[t];
+    int64_t run = v - s + (w > 0 ? wsum[w - 1] : 0);
+    if (t == (int)blockDim.x - 1) offsets[k] = run + s;
     for (int j = lo; j < hi; ++j) {
         offsets[j] = run;
         run += counts[j];
