@@ -457,11 +457,31 @@ def run_ours(args):
         host_ms.clear()
         if world > 1:
             dist.barrier()
-        ems = e2e_run(e2e_steps)
+        def timed_e2e():
+            t_ms = e2e_run(e2e_steps)
+            if world > 1:
+                t = torch.tensor([t_ms], device=dev, dtype=torch.float64)
+                dist.all_reduce(t, op=dist.ReduceOp.MAX)
+                t_ms = float(t.item())
+            return t_ms
+
+        ems = timed_e2e()
+        # The host link is shared with the host's other traffic: a run whose
+        # copies averaged under 3/4 of the rate probed just before it is taken
+        # again once (both attempts are reported).
+        probe = h2d_probe_gbs
         if world > 1:
-            t = torch.tensor([ems], device=dev, dtype=torch.float64)
-            dist.all_reduce(t, op=dist.ReduceOp.MAX)
-            ems = float(t.item())
+            t = torch.tensor([probe], device=dev, dtype=torch.float64)
+            dist.all_reduce(t, op=dist.ReduceOp.MIN)
+            probe = float(t.item())
+        first_attempt = None
+        if h2d / (ems / e2e_steps / 1e3) / 1e9 < 0.75 * probe:
+            first_attempt = {"ms_per_step": ems / e2e_steps,
+                             "h2d_effective_gbs": round(h2d / (ems / e2e_steps / 1e3) / 1e9, 1)}
+            host_ms.clear()
+            if world > 1:
+                dist.barrier()
+            ems = timed_e2e()
         # and right after it: the link is shared with the host's other traffic
         torch.cuda.synchronize()
         p0.record(stream)
@@ -474,6 +494,7 @@ def run_ours(args):
                "host_enqueue_ms_per_step": round(statistics.mean(host_ms), 3),
                "h2d_probe_gbs": round(h2d_probe_gbs, 1), "h2d_probe_after_gbs": round(h2d_probe_after_gbs, 1),
                "h2d_effective_gbs": round(h2d / (ems / e2e_steps / 1e3) / 1e9, 1),
+               "remeasured_after": first_attempt,
                "ms_per_step": ems / e2e_steps,
                "path": f"pinned host fp32 points -> H2D in {nchunk} row ranges on a copy stream (two device "
                        "buffers: the next step's points stream in during this step's tail), each range assigned "
