@@ -218,7 +218,9 @@ int skm_pca_fit(const float *X, int64_t n, int d, int d_out, float *mean, float 
  *  repr = SKM_REPR_RBQ1 (RabitQ, 1-bit): mean m (fp64 sum, rounded to fp32)
  *    when fit != 0, else the supplied m; r = x - m; bit i = (r_i > 0);
  *    nx2 = ||r||^2; F = sqrt(d) ||r||^2 / ||r||_1 (0 when r = 0), i.e.
- *    ||r|| / <xbar, x>; popx = set bits.  Outputs: codes uint32[n][W],
+ *    ||r|| / <xbar, x>; popx = set bits.  nx2 and F come from compensated
+ *    fp32 sums: within about 5 x 2^-24 and 12 x 2^-24 relative of the exact
+ *    values (the bits are exact).  Outputs: codes uint32[n][W],
  *    W = ceil(d/32), bit j of word w = dim 32w+j (unused high bits are 0);
  *    nx2, F float[n]; popx int32[n]; m float[d].
  *  repr = SKM_REPR_LVQ4 (Section 3.1 "LVQ4", per-vector): b = min_i x_i,
