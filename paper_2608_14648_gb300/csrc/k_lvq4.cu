@@ -396,12 +396,11 @@ __global__ void __launch_bounds__(256) assign_lvq4_simt_kernel(const uint32_t *_
 __global__ void lvq4_q_kernel(const float4 *__restrict__ fac, const int32_t *__restrict__ perm,
                               const int64_t *__restrict__ offsets, int k, int e, uint32_t *__restrict__ sq,
                               int64_t *__restrict__ bq) {
-    const double pow2 = ldexp(1.0, e);
     const int64_t nval = offsets[k];
     for (int64_t q = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; q < nval; q += (int64_t)gridDim.x * blockDim.x) {
         const float4 f = fac[perm[q]];
-        sq[q] = (uint32_t)__double2ll_rn(__dmul_rn((double)f.x, pow2));
-        bq[q] = __double2ll_rn(__dmul_rn((double)f.y, pow2));
+        sq[q] = (uint32_t)fixed_rint(f.x, e);
+        bq[q] = fixed_rint(f.y, e);
     }
 }
 

@@ -300,11 +300,10 @@ __device__ __forceinline__ float rbq1_finish(int64_t T, int64_t U, float m, doub
 __global__ void rbq1_fq_kernel(const float *__restrict__ F, const int32_t *__restrict__ perm,
                                const int64_t *__restrict__ offsets, int k, int e,
                                int64_t *__restrict__ fq) {
-    const double pow2 = ldexp(1.0, e);
     const int64_t nval = offsets[k];
     for (int64_t q = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; q < nval;
          q += (int64_t)gridDim.x * blockDim.x)
-        fq[q] = __double2ll_rn(__dmul_rn((double)F[perm[q]], pow2));
+        fq[q] = fixed_rint(F[perm[q]], e);
 }
 
 cudaError_t launch_rbq1_fq(const float *F, const int32_t *perm, const int64_t *offsets, int k,

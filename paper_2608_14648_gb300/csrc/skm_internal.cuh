@@ -55,6 +55,36 @@ struct Carver {
 inline int words_of(int d) { return (d + 31) / 32; }
 inline int64_t cdiv(int64_t a, int64_t b) { return (a + b - 1) / b; }
 
+// rint(v 2^e) as an integer, rounding half to even, for a finite v and
+// |v 2^e| < 2^62: v's 24-bit significand is shifted by its exponent plus e and
+// the dropped bits are rounded in integer arithmetic, so the result equals the
+// exact fp64 product rounded to an integer, without fp64 instructions (which
+// GB300 issues at a small fraction of the integer rate).
+__device__ __forceinline__ int64_t fixed_rint(float v, int e) {
+    const uint32_t b = __float_as_uint(v);
+    const int E = (int)((b >> 23) & 0xffu);
+    uint64_t m = b & 0x7fffffu;
+    int sh;
+    if (E) {
+        m |= 0x800000u;
+        sh = E - 150 + e;
+    } else {
+        sh = -149 + e;
+    }
+    uint64_t q;
+    if (sh >= 0) {
+        q = m << sh;
+    } else if (-sh > 25) {  // m < 2^24: below one half
+        q = 0;
+    } else {
+        const int s = -sh;
+        q = m >> s;
+        const uint64_t r = m & ((1ull << s) - 1ull), half = 1ull << (s - 1);
+        if (r > half || (r == half && (q & 1ull))) ++q;
+    }
+    return (b >> 31) ? -(int64_t)q : (int64_t)q;
+}
+
 // acc += f when (word & mask) != 0: one bit test and one predicated 32-bit add
 // (the 1-bit decode-average sums of a run of rows).
 __device__ __forceinline__ void add_if_bit(uint32_t &acc, uint32_t word, uint32_t mask, uint32_t f) {
