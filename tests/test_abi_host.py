@@ -150,3 +150,14 @@ def test_symmetric_flag_is_validated(skm):
     r = skm.Data(skm.REPR_RBQ1, 16, 100, 0x1000, FAKE, FAKE, FAKE, FAKE, 0, skm.FLAG_SYMMETRIC)
     assert L.skm_assign_rbq1_noalloc(ctypes.byref(r), FAKE, 4, FAKE, None, None) == 2
     assert L.skm_workspace_size(0, ctypes.byref(r), 4) > 0
+
+
+def test_copy_from_host_arguments(skm):
+    L = skm.lib()
+    FAKE = ctypes.c_void_p(0x1000)
+    # zero bytes: a no-op that touches nothing
+    assert L.skm_copy_from_host(None, None, 0, None) == 0
+    # NULL destination or source with bytes to copy: rejected before any CUDA call
+    assert L.skm_copy_from_host(None, FAKE, 16, None) == 1
+    assert L.skm_copy_from_host(FAKE, None, 16, None) == 1
+    assert "NULL" in L.skm_last_error().decode()
