@@ -335,7 +335,10 @@ int skm_assign(const skm_data *x, const void *C, int k, const int32_t *prev_assi
  *   (nothing is launched).
  *   The first call on a device looks up the array's device address with that
  *   device current (cudaGetSymbolAddress) and caches it; make that first call
- *   before any stream capture.
+ *   before any stream capture.  The cached address belongs to the device's
+ *   current (primary) context: do not use this entry point across a
+ *   cudaDeviceReset or anything else that destroys and recreates that context,
+ *   because the array then moves and the cached address goes stale.
  *   All calls share the array and it keeps the last call's contents: calls
  *   whose work overlaps on the GPU (other streams, other threads) race; order
  *   them on one stream or synchronise between them.

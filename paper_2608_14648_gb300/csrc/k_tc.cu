@@ -56,15 +56,9 @@ constexpr int TCAND = 4;
 constexpr unsigned long long WAIT_LIMIT_NS = 2000000000ull;  // 2 s per barrier wait
 
 enum { MODE_SCREEN = 0, MODE_SQ8 = 1, MODE_RBQ1 = 2, MODE_LVQ4 = 3, MODE_GEMM = 4 };
-// epilogue warps per TMEM lane quarter, and CTAs per cluster (centroid
-// slices multicast across the cluster), by mode.  Clusters of 2 run
-// correctly but measured slower on GB300 (the pair's pipelines wait on each
-// other's slowest epilogue: fp32 0.999 vs 0.956 ms, 1-bit 0.602 vs 0.554 ms
-// at 1M x 1000 x 768 with one job stream; with two job streams 1-bit 0.516
-// vs 0.512 ms, LVQ4 0.537 vs 0.516 ms), so every mode runs one CTA per
-// cluster.  Segmented mode always does.
+// Epilogue warps per TMEM lane quarter, by mode.  Every CTA works alone
+// (no thread-block clusters): it loads its own centroid slices.
 constexpr int TC_NH[5] = {4, 4, 4, 4, 4};
-constexpr int TC_CL[5] = {1, 1, 1, 1, 1};
 // Job streams per CTA, by mode.  NS = 2: the CTA's point tiles form two
 // streams whose jobs the MMA warp issues alternately, each into its own TMEM
 // accumulator, each drained by its own half of the epilogue warps; an
@@ -211,37 +205,6 @@ __device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap *map
         "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(bar)
         : "memory");
 }
-// Multicast form: the box lands at the same shared-memory offset in every CTA
-// of the cluster named in `mask`, and each of their mbarriers at `bar`
-// receives the completed bytes.
-__device__ __forceinline__ void tma_load_2d_mc(uint32_t dst, const CUtensorMap *map, int x, int y,
-                                               uint32_t bar, uint16_t mask) {
-    asm volatile(
-        "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes.multicast::cluster"
-        " [%0], [%1, {%2, %3}], [%4], %5;" ::"r"(dst),
-        "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(bar), "h"(mask)
-        : "memory");
-}
-__device__ __forceinline__ uint32_t cluster_rank() {
-    uint32_t r;
-    asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
-    return r;
-}
-__device__ __forceinline__ uint32_t cluster_index() {
-    uint32_t r;
-    asm volatile("mov.u32 %0, %%clusterid.x;" : "=r"(r));
-    return r;
-}
-__device__ __forceinline__ uint32_t cluster_count() {
-    uint32_t r;
-    asm volatile("mov.u32 %0, %%nclusterid.x;" : "=r"(r));
-    return r;
-}
-// every thread of every CTA of the cluster
-__device__ __forceinline__ void cluster_sync_all() {
-    asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" ::
-                     : "memory");
-}
 __device__ __forceinline__ void tc_fence_before() {
     asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
 }
@@ -252,15 +215,6 @@ __device__ __forceinline__ void tc_commit(uint32_t bar) {
     asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(
                      bar)
                  : "memory");
-}
-// arrive on the mbarrier at `bar` in every CTA of the cluster named in `mask`
-// once the MMAs issued so far have completed
-__device__ __forceinline__ void tc_commit_mc(uint32_t bar, uint16_t mask) {
-    asm volatile(
-        "tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64 [%0], %1;" ::"r"(
-            bar),
-        "h"(mask)
-        : "memory");
 }
 __device__ __forceinline__ void tc_mma(uint32_t dtmem, uint64_t adesc, uint64_t bdesc, uint32_t idesc,
                                        uint32_t accumulate) {
@@ -454,12 +408,11 @@ __device__ __forceinline__ void ct_range(const TcParams &p, int64_t rt, int &lo,
     }
 }
 
-template <int MODE, int NH, int CL, bool SEG, int NS>
+template <int MODE, int NH, bool SEG, int NS>
 __global__ void __launch_bounds__(tc_threads<NH>(), 1)
     tc_assign_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                      const TcParams p) {
     static_assert(NS == 1 || (NS == 2 && NH % 2 == 0), "two job streams: two epilogue groups");
-    static_assert(CL == 1 || !SEG, "segmented mode: one CTA per cluster");
     static_assert(NS == 1 || MODE == MODE_GEMM || epi_threads<NH>() / NS >= (MODE == MODE_SCREEN ? 128 : 256),
                   "records staged by one epilogue group");
     extern __shared__ uint8_t smem_raw[];
@@ -485,7 +438,7 @@ __global__ void __launch_bounds__(tc_threads<NH>(), 1)
     if (threadIdx.x == 0) {
         for (int s = 0; s < STAGES; ++s) {
             mbar_init(full_bar(s), 1);
-            mbar_init(empty_bar(s), CL);  // one MMA commit per CTA of the cluster
+            mbar_init(empty_bar(s), 1);  // the MMA warp's commit
         }
         for (int b = 0; b < 2; ++b) {
             mbar_init(tfull_bar(b), 1);
@@ -506,18 +459,10 @@ __global__ void __launch_bounds__(tc_threads<NH>(), 1)
     __syncthreads();
     tc_fence_after();
     const uint32_t tmem = *tmem_slot;
-    // Cluster of CL CTAs: they walk the point tiles in lockstep (CTA r of
-    // cluster c takes point tile (c + i nclusters) CL + r) over the same
-    // centroid tiles, and each loads 256 / CL rows of every centroid slice
-    // with multicast into all of them, so a slice leaves L2 once per cluster.
-    // A stage is free again once every CTA's MMAs have read it (empty
-    // barriers count CL commits).  A tile index past the last point tile
-    // loads zeros (TMA out-of-range fill) and writes nothing.
-    const uint32_t crank = CL > 1 ? cluster_rank() : 0u;
-    const int64_t g0 = CL > 1 ? (int64_t)cluster_index() : (int64_t)blockIdx.x;
-    const int64_t gstep = CL > 1 ? (int64_t)cluster_count() : (int64_t)gridDim.x;
-    const int64_t ngroups = (p.nrt + CL - 1) / CL;
-    if (CL > 1) cluster_sync_all();  // peers' barriers are initialised before any multicast
+    // CTA b takes the point tiles b, b + grid, b + 2 grid, ...
+    const int64_t g0 = (int64_t)blockIdx.x;
+    const int64_t gstep = (int64_t)gridDim.x;
+    const int64_t ngroups = p.nrt;
 
     // Job order (producer and MMA issuer walk it identically): stream s takes
     // the CTA's point-tile groups g0 + (s + NS i) gstep; the streams' jobs
@@ -529,7 +474,7 @@ __global__ void __launch_bounds__(tc_threads<NH>(), 1)
     auto stream_seek = [&](JobStream &js) {  // the first job at or after group js.g
         while (js.g < ngroups) {
             int lo, hi;
-            ct_range(p, js.g * CL + crank, lo, hi);
+            ct_range(p, js.g, lo, hi);
             if (lo < hi) {
                 js.ct = lo;
                 js.hi = hi;
@@ -578,7 +523,7 @@ __global__ void __launch_bounds__(tc_threads<NH>(), 1)
                 int64_t gj;
                 int ct;
                 stream_take(js, sj, gj, ct);
-                const int64_t rt = gj * CL + crank;
+                const int64_t rt = gj;
                 turn = (sj + 1) % NS;
                 {
                     for (int kt = 0; kt < NSEG * p.nkc; ++kt, ++it) {
@@ -589,12 +534,7 @@ __global__ void __launch_bounds__(tc_threads<NH>(), 1)
                         if (!mbar_wait(empty_bar(s), ph ^ 1u, abort_flag)) goto producer_done;
                         mbar_expect_tx(full_bar(s), A_STAGE + B_STAGE);
                         tma_load_2d(sA + s * A_STAGE, &tmA, kc * KC_ELEMS, arow, full_bar(s));
-                        if (CL == 1)
-                            tma_load_2d(sB + s * B_STAGE, &tmB, kc * KC_ELEMS, brow, full_bar(s));
-                        else
-                            tma_load_2d_mc(sB + s * B_STAGE + crank * (B_STAGE / CL), &tmB, kc * KC_ELEMS,
-                                           ct * BN + (int)crank * (BN / CL), full_bar(s),
-                                           (uint16_t)((1u << CL) - 1u));
+                        tma_load_2d(sB + s * B_STAGE, &tmB, kc * KC_ELEMS, brow, full_bar(s));
                     }
                 }
             }
@@ -640,10 +580,7 @@ __global__ void __launch_bounds__(tc_threads<NH>(), 1)
                             else
                                 tc_mma(dcol, ad + 2u * kk, bd + 2u * kk, IDESC, (kc | kk) != 0);
                         }
-                        if (CL == 1)
-                            tc_commit(empty_bar(s));
-                        else
-                            tc_commit_mc(empty_bar(s), (uint16_t)((1u << CL) - 1u));
+                        tc_commit(empty_bar(s));
                     }
                     tc_commit(tfull_bar(b));
                 }
@@ -700,7 +637,7 @@ __global__ void __launch_bounds__(tc_threads<NH>(), 1)
         };
         {
             int lo0, hi0;
-            ct_range(p, (g0 + grp * gstep) * CL + crank, lo0, hi0);
+            ct_range(p, g0 + grp * gstep, lo0, hi0);
             rec_load(lo0);
         }
         // A warp whose barrier wait gave up stops computing but keeps taking part
@@ -708,7 +645,7 @@ __global__ void __launch_bounds__(tc_threads<NH>(), 1)
         bool dead = false;
         uint32_t job = 0;  // jobs of this group so far (NS = 1: of the CTA)
         for (int64_t g = g0 + grp * gstep; g < ngroups; g += NS * gstep) {
-            const int64_t rt = g * CL + crank;
+            const int64_t rt = g;
             const int64_t row = rt * BM + rin;
             const bool valid = row < p.n;
             ScreenRow sr;
@@ -730,7 +667,7 @@ __global__ void __launch_bounds__(tc_threads<NH>(), 1)
             int next_lo = 0;
             {
                 int nhi;
-                ct_range(p, (g + NS * gstep) * CL + crank, next_lo, nhi);
+                ct_range(p, g + NS * gstep, next_lo, nhi);
             }
             if (MODE == MODE_SCREEN) {
                 a2 = valid ? 2.0f * p.xinfo[row].x : 0.0f;
@@ -1119,9 +1056,6 @@ __global__ void __launch_bounds__(tc_threads<NH>(), 1)
     }
     tc_fence_before();
     __syncthreads();
-    // no CTA leaves while a peer may still multicast into its shared memory
-    // or arrive on its barriers
-    if (CL > 1) cluster_sync_all();
     if (warp == 1) {
         __syncwarp();
         tc_fence_after();
@@ -1549,58 +1483,39 @@ int device_sms() {
     return sms > 0 ? sms : 148;
 }
 
-// Segmented mode runs one CTA per cluster: the CTAs of a cluster would walk
-// different centroid ranges, so there is no common slice to multicast.
-template <int MODE, int CL, bool SEG>
-int launch_tc_cl(const void *xs, int64_t n, int dp, int d, const void *cs, int k, const TcParams &p0,
-                 cudaStream_t st);
+template <int MODE, bool SEG>
+int launch_tc_kind(const void *xs, int64_t n, int dp, int d, const void *cs, int k, const TcParams &p0,
+                   cudaStream_t st);
 
 template <int MODE>
 int launch_tc(const void *xs, int64_t n, int dp, int d, const void *cs, int k, const TcParams &p0,
               cudaStream_t st) {
-    if (p0.seg_group) return launch_tc_cl<MODE, 1, true>(xs, n, dp, d, cs, k, p0, st);
-    return launch_tc_cl<MODE, TC_CL[MODE], false>(xs, n, dp, d, cs, k, p0, st);
+    if (p0.seg_group) return launch_tc_kind<MODE, true>(xs, n, dp, d, cs, k, p0, st);
+    return launch_tc_kind<MODE, false>(xs, n, dp, d, cs, k, p0, st);
 }
 
-template <int MODE, int CL, bool SEG>
-int launch_tc_cl(const void *xs, int64_t n, int dp, int d, const void *cs, int k, const TcParams &p0,
-                 cudaStream_t st) {
+// One persistent CTA per SM (at most one point tile per CTA when there are
+// fewer tiles than SMs).
+template <int MODE, bool SEG>
+int launch_tc_kind(const void *xs, int64_t n, int dp, int d, const void *cs, int k, const TcParams &p0,
+                   cudaStream_t st) {
     constexpr int NH = TC_NH[MODE];
     constexpr int NS = TC_NS[MODE];
     constexpr size_t SMEM = tc_smem_bytes<MODE, NH, NS>();
     static_assert(SMEM <= 227 * 1024, "shared memory per CTA");
-    auto kern = tc_assign_kernel<MODE, NH, CL, SEG, NS>;
+    auto kern = tc_assign_kernel<MODE, NH, SEG, NS>;
     const int segi = SEG ? 1 : 0;
-    // per device: the attribute and the number of clusters that fit at once
+    // the dynamic shared memory attribute, set once per device
     constexpr int MAXDEV = 64;
     static std::mutex mu;
-    static int cached_clusters[5][2][MAXDEV] = {};
+    static bool attr_set[5][2][MAXDEV] = {};
     int dev = 0;
     SKM_CUDA_TRY(cudaGetDevice(&dev));
-    int max_clusters = 0;
     {
         std::lock_guard<std::mutex> lock(mu);
-        if (dev < MAXDEV) max_clusters = cached_clusters[MODE][segi][dev];
-        if (max_clusters == 0) {
+        if (dev >= MAXDEV || !attr_set[MODE][segi][dev]) {
             SKM_CUDA_TRY(cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)SMEM));
-            if (CL > 1) {
-                cudaLaunchConfig_t qc = {};
-                qc.gridDim = dim3((unsigned)(CL * device_sms()));
-                qc.blockDim = dim3(tc_threads<NH>());
-                qc.dynamicSmemBytes = SMEM;
-                cudaLaunchAttribute qa[1];
-                qa[0].id = cudaLaunchAttributeClusterDimension;
-                qa[0].val.clusterDim.x = CL;
-                qa[0].val.clusterDim.y = 1;
-                qa[0].val.clusterDim.z = 1;
-                qc.attrs = qa;
-                qc.numAttrs = 1;
-                SKM_CUDA_TRY(cudaOccupancyMaxActiveClusters(&max_clusters, kern, &qc));
-            } else {
-                max_clusters = device_sms();
-            }
-            if (max_clusters < 1) return set_error(SKM_ERR_CUDA, "no cluster of %d CTAs fits on this device", CL);
-            if (dev < MAXDEV) cached_clusters[MODE][segi][dev] = max_clusters;
+            if (dev < MAXDEV) attr_set[MODE][segi][dev] = true;
         }
     }
     CUtensorMap ma, mb;
@@ -1608,28 +1523,15 @@ int launch_tc_cl(const void *xs, int64_t n, int dp, int d, const void *cs, int k
     // GEMM mode: the A and B parts are stacked (rows [part][n], [part][k])
     const int parts = MODE == MODE_GEMM ? 3 : 1;
     SKM_TRY(make_map(&ma, xs, parts * n, d, dp, BM, eb));
-    SKM_TRY(make_map(&mb, cs, (int64_t)parts * k, d, dp, BN / CL, eb));
+    SKM_TRY(make_map(&mb, cs, (int64_t)parts * k, d, dp, BN, eb));
     TcParams p = p0;
     p.n = n;
     p.nrt = cdiv(n, BM);
     p.k = k;
     p.nct = (int)cdiv(k, BN);
     p.nkc = (int)cdiv(d, 128 / eb);
-    const int64_t groups = cdiv(p.nrt, CL);
-    const int grid = CL * (int)std::min<int64_t>(max_clusters, groups);
-    cudaLaunchConfig_t cfg = {};
-    cfg.gridDim = dim3((unsigned)grid);
-    cfg.blockDim = dim3(tc_threads<NH>());
-    cfg.dynamicSmemBytes = SMEM;
-    cfg.stream = st;
-    cudaLaunchAttribute attr[1];
-    attr[0].id = cudaLaunchAttributeClusterDimension;
-    attr[0].val.clusterDim.x = CL;
-    attr[0].val.clusterDim.y = 1;
-    attr[0].val.clusterDim.z = 1;
-    cfg.attrs = attr;
-    cfg.numAttrs = 1;
-    SKM_CUDA_TRY(cudaLaunchKernelEx(&cfg, kern, ma, mb, p));
+    const int grid = (int)std::min<int64_t>(device_sms(), p.nrt);
+    kern<<<grid, tc_threads<NH>(), SMEM, st>>>(ma, mb, p);
     SKM_CUDA_TRY(launched());
     return SKM_OK;
 }
