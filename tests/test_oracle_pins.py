@@ -756,3 +756,139 @@ def test_rbq1_symmetric_exact_for_sign_constant_vectors():
     D = cdist(X.astype(np.float64), C.astype(np.float64), "sqeuclidean")
     np.testing.assert_allclose(est, D[np.arange(n), a], rtol=1e-5)
     np.testing.assert_array_equal(a, D.argmin(1))
+
+
+# ------------------------------------- hierarchical SQ8 / RBQ1, bf16 update and objective
+def test_hierarchical_sq8_with_one_meso_cluster_is_plain_lloyd():
+    """m = 1: the fine phase is plain SQ8 Lloyd (pinned against exact integer
+    means above) from the evenly spaced members floor(t n / k)."""
+    r = _rng(51)
+    n, d, k = 500, 12, 7
+    codes = r.integers(0, 256, (n, d)).astype(np.uint8)
+    C, a, am, kf = oracle.hierarchical("sq8", codes, k, 1, np.array([4]), 2, 4)
+    assert kf == [k] and np.all(am == 0)
+    init = np.array(oracle.fine_init_positions(n, k))
+    Cl, al = oracle.lloyd_sq8(codes, codes[init], 4)
+    np.testing.assert_array_equal(a, al)
+    np.testing.assert_array_equal(C, Cl)
+
+
+def test_hierarchical_rbq1_with_one_meso_cluster_is_plain_lloyd():
+    """m = 1: the fine phase is plain RabitQ Lloyd from the decoded evenly
+    spaced members."""
+    r = _rng(52)
+    n, d, k = 400, 40, 5
+    X = r.standard_normal((n, d)).astype(np.float32)
+    m = oracle.rbq1_mean(X)
+    codes, nx2, F, popx = oracle.rbq1_encode(X, m)
+    e = oracle.rbq1_exponent(F)
+    data = {"codes": codes, "nx2": nx2, "F": F, "popx": popx, "d": d, "m": m, "e": e}
+    C, a, am, kf = oracle.hierarchical("rbq1", data, k, 1, np.array([7]), 2, 3)
+    assert kf == [k] and np.all(am == 0)
+    init = np.array(oracle.fine_init_positions(n, k))
+    C0 = oracle.rbq1_decode_points(codes, F, d, m, e, init)
+    Cl, al = oracle.lloyd_rbq1(codes, nx2, F, popx, d, m, C0, 3, e)
+    np.testing.assert_array_equal(a, al)
+    np.testing.assert_array_equal(C, Cl)
+
+
+def _blobs(r, d, sep, sub, noise, per=50):
+    """Four far-apart blobs of three sub-blobs each (labels 0..11 in order):
+    blob centres sep * e_b, sub-blob offsets sub * e_{4 + s} along axes of
+    their own, isotropic Gaussian noise."""
+    pts, labels = [], []
+    for b in range(4):
+        for s in range(3):
+            c = np.zeros(d)
+            c[b] = sep
+            c[4 + 3 * b + s] = sub
+            pts.append(c + r.normal(0, noise, (per, d)))
+            labels.append(np.full(per, 3 * b + s))
+    return np.concatenate(pts).astype(np.float32), np.concatenate(labels)
+
+
+def _assert_blobs_recovered(a, am, kf, labels):
+    assert kf == [3, 3, 3, 3]
+    for b in range(4):  # each blob is one meso cluster
+        assert len(set(am[labels // 3 == b])) == 1
+    for s in range(12):  # each sub-blob is one fine cluster, and they are distinct
+        assert len(set(a[labels == s])) == 1
+    assert len({int(a[labels == s][0]) for s in range(12)}) == 12
+
+
+def test_hierarchical_sq8_recovers_separated_blobs():
+    """SQ8 codes of four far-apart blobs of three sub-blobs each, m = 4 meso
+    and k = 12 fine clusters: meso clusters are the blobs (3 fine clusters
+    each), fine clusters the sub-blobs."""
+    r = _rng(53)
+    X, labels = _blobs(r, 16, 100.0, 20.0, 0.5)
+    b, s = oracle.sq8_fit(X)
+    codes = oracle.sq8_encode(X, b, s)
+    meso_init = np.array([0, 150, 300, 450])
+    C, a, am, kf = oracle.hierarchical("sq8", codes, 12, 4, meso_init, 3, 5)
+    _assert_blobs_recovered(a, am, kf, labels)
+    C2, a2, _, _ = oracle.hierarchical("sq8", codes, 12, 4, meso_init, 3, 5, refine=True)
+    np.testing.assert_array_equal(a2, a)  # a fixed point: refinement changes nothing
+
+
+def _sign_blobs(r, per=50):
+    """Four blobs of three sub-blobs each (labels 0..11 in order) for 1-bit
+    codes, which see only the signs of x - m: on dimensions 0..31 each blob
+    has a +-30 pattern (every dimension + for two blobs and - for the other
+    two, so the data mean is 0 there), on dimensions 32..63 each sub-blob a
+    pattern of +10, -10 and 0 (a permutation per blob and dimension, mean 0),
+    plus Gaussian noise 0.5.  Blobs are then ~8x farther apart than
+    sub-blobs, and every blob and sub-blob has a sign code of its own."""
+    pats = [(1, 1, -1, -1), (1, -1, 1, -1), (1, -1, -1, 1), (-1, -1, 1, 1), (-1, 1, -1, 1), (-1, 1, 1, -1)]
+    B = np.array([pats[r.integers(0, 6)] for _ in range(32)], np.float64).T * 30.0  # [4][32]
+    S = np.zeros((4, 3, 32))
+    for b in range(4):
+        for i in range(32):
+            S[b, :, i] = r.permutation([10.0, -10.0, 0.0])
+    pts, labels = [], []
+    for b in range(4):
+        for s in range(3):
+            c = np.concatenate([B[b], S[b, s]])
+            pts.append(c + r.normal(0, 0.5, (per, 64)))
+            labels.append(np.full(per, 3 * b + s))
+    return np.concatenate(pts).astype(np.float32), np.concatenate(labels)
+
+
+def test_hierarchical_rbq1_recovers_separated_blobs():
+    """Blobs and sub-blobs with sign codes of their own, as RabitQ 1-bit
+    codes (d = 64), m = 4 meso and k = 12 fine clusters: meso clusters are
+    the blobs, fine clusters the sub-blobs."""
+    r = _rng(54)
+    X, labels = _sign_blobs(r)
+    m = oracle.rbq1_mean(X)
+    codes, nx2, F, popx = oracle.rbq1_encode(X, m)
+    e = oracle.rbq1_exponent(F)
+    data = {"codes": codes, "nx2": nx2, "F": F, "popx": popx, "d": 64, "m": m, "e": e}
+    meso_init = np.array([0, 150, 300, 450])
+    C, a, am, kf = oracle.hierarchical("rbq1", data, 12, 4, meso_init, 3, 5)
+    _assert_blobs_recovered(a, am, kf, labels)
+
+
+def test_update_bf16_is_member_mean_of_decoded_rows_and_keeps_empty():
+    r = _rng(55)
+    n, d, k = 300, 21, 6
+    Xb = oracle.round_bf16(r.standard_normal((n, d)))
+    Xf = oracle.bf16_to_f32(Xb).astype(np.float64)
+    a = r.integers(0, k - 1, n).astype(np.int32)  # cluster k-1 stays empty
+    C0 = r.standard_normal((k, d)).astype(np.float32)
+    C, counts = oracle.update_bf16(Xb, a, C0)
+    np.testing.assert_array_equal(counts, np.bincount(a, minlength=k))
+    for j in range(k - 1):
+        np.testing.assert_allclose(C[j], Xf[a == j].mean(axis=0), rtol=1e-6, atol=1e-7)
+    np.testing.assert_array_equal(C[k - 1], C0[k - 1])
+
+
+def test_objective_bf16_is_wcss_of_decoded_rows():
+    r = _rng(56)
+    n, d, k = 120, 19, 5
+    Xb = oracle.round_bf16(r.standard_normal((n, d)))
+    C = r.standard_normal((k, d)).astype(np.float32)
+    a = r.integers(0, k, n).astype(np.int32)
+    D = cdist(oracle.bf16_to_f32(Xb).astype(np.float64), C.astype(np.float64), "sqeuclidean")
+    want = float(D[np.arange(n), a].sum())
+    assert math.isclose(oracle.objective_bf16(Xb, C, a), want, rel_tol=1e-12)
