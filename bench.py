@@ -1,19 +1,23 @@
 #!/usr/bin/env python
 """Benchmark of the Lloyd k-means hot path on GB300.
 
-Workload: 1,000,000 unit-norm synthetic embeddings, d = 768 (2,000-component
-Gaussian mixture, per-dimension variance (1+j)^-0.5, Haar rotation, L2
-normalisation), k = 1,000, clustered both as raw fp32 and as RabitQ 1-bit
-codes.  One step = one Lloyd iteration (assign + update) of each
-representation, i.e. 2 * N * k point-centroid distances.  Metric:
-point-centroid distances per second per Lloyd iteration.
+Headline workload (emb10m_pca256): 10,000,000 unit-norm synthetic embeddings,
+D = 1024 (10,000-component Gaussian mixture, per-dimension variance
+(1+j)^-0.5, Haar rotation, L2 normalisation), PCA-projected to d' = 256 (fp32
+projection, bf16 storage), k = 10,000.  One step = one Lloyd iteration (STEP 2
+assignment + STEP 3 update) over all points, i.e. N * k point-centroid
+distances.  Metric: point-centroid distances per second per Lloyd iteration.
+Beside it the line reports the 1M x 768 (fp32 and 1-bit) and 10M x 1024
+(1-bit, k = 3,162) iterations, the pruned assignment of the headline
+workload, and the end-to-end step from pinned host memory.
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
 
 N > 1 runs under torchrun, one rank per GPU: every rank clusters its own
-1M-point shard (weak scaling) and the update's cluster sums and counts are
-all-reduced once per representation per step (the path's one exchange).
---impl reference times the CPU oracle on a bounded sample of the workload.
+10M-point shard (weak scaling); the PCA basis and the initial centroids come
+from rank 0, and the update's cluster sums and counts are all-reduced once per
+step (the path's one exchange).  --impl reference times the CPU oracle on a
+bounded sample of the headline workload.
 """
 from __future__ import annotations
 
@@ -29,19 +33,24 @@ import time
 ROOT = os.path.dirname(os.path.abspath(__file__))
 sys.path.insert(0, ROOT)
 
-N_POINTS, DIM, K, N_COMP = 1_000_000, 768, 1000, 2000
+HEAD = "emb10m_pca256"
+D_PCA = 256
 METRIC = "k-means point·centroid distances/s per Lloyd iter (1 GB300); % of roofline"
-WORKLOAD = "emb1m_d768: N=1,000,000 x d=768 unit-norm GMM embeddings, k=1,000; fp32 + RabitQ 1-bit"
+WORKLOAD = ("emb10m_pca256: N=10,000,000 unit-norm GMM embeddings, D=1024 -> PCA d'=256 (fp32 projection, "
+            "bf16 storage), k=10,000")
 SM_COUNT = 152
 # row ranges of the end-to-end step's host-to-device copy (overlapped with work)
 E2E_CHUNKS = 16
 # POPC results per clock per SM used for the 1-bit kernel's ALU roofline
 # (measured 15.9 on GB300 with a throughput probe).
 POPC_PER_CLK_SM = 16
-# DRAM bytes (read + write) per point of the assignment kernels, from one ncu
-# capture each (200,000 points x d=768, k=1000; profiles/tc_assign_*.md).
-# Each point row is read once per launch, so traffic scales with the points.
+# DRAM bytes (read + write) per point of the assignment kernels, each from
+# one ncu capture of a smaller case of the same kernel (every point row is
+# read once per launch, so traffic scales with the points): the bf16 screen
+# at 400,000 x 256 with k = 10,000; the fp32 screen and the e4m3 1-bit
+# kernel at 200,000 x 768 with k = 1,000.
 TRAFFIC_PER_POINT = {
+    "assign_bf16_screen": (213.449216e6 + 4.711680e6) / 400_000,
     "assign_f32": (314.849280e6 + 5.701888e6) / 200_000,
     "assign_rbq1": (156.890624e6 + 3.590912e6) / 200_000,
 }
@@ -124,24 +133,220 @@ class ClockSampler:
 
 
 # ----------------------------------------------------------------------------
-def cpu_baseline_sample(X_host, C32, codes, nx2, F, popx, m, e, Cr, budget_s=12.0):
-    """Oracle (as it stands) on a bounded row sample: one Lloyd iteration of
-    each representation.  Returns (distances/s, rows, seconds, threads)."""
+def _graph_of(step, stream):
+    """Captures step() once in a CUDA graph (after one run on a side stream);
+    returns (graph, library launches per step) or (None, note)."""
+    import torch
+
+    import paper_2608_14648_gb300 as skm
+
+    try:
+        side = torch.cuda.Stream()
+        side.wait_stream(stream)
+        with torch.cuda.stream(side):
+            step()
+        stream.wait_stream(side)
+        torch.cuda.synchronize()
+        l0 = skm.skm_kernel_launches()
+        graph = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(graph):
+            step()
+        launches = skm.skm_kernel_launches() - l0
+        graph.replay()
+        torch.cuda.synchronize()
+        return graph, launches
+    except Exception as exc:  # eager steps instead, reported
+        return None, f"graph capture failed, eager steps: {exc!r}"[:200]
+
+
+def _timed_steps(step, stream, steps, warmup, world, dist, local_rank, use_graph):
+    """warmup eager steps, then `steps` steps (CUDA-graph replays on one GPU)
+    bracketed by a barrier and synchronisation; returns (ms max over ranks,
+    launches, timing note, clocks)."""
+    import torch
+
+    import paper_2608_14648_gb300 as skm
+
+    for _ in range(warmup):
+        step()
+    torch.cuda.synchronize()
+    graph, lps, note = None, None, None
+    if use_graph:
+        graph, lps = _graph_of(step, stream)
+        if graph is None:
+            note, lps = lps, None
+    if world > 1:
+        dist.barrier()
+    clocks = ClockSampler(local_rank)
+    clocks.start()
+    torch.cuda.synchronize()
+    l0 = skm.skm_kernel_launches()
+    t0, t1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    t0.record(stream)
+    for _ in range(steps):
+        if graph is not None:
+            graph.replay()
+        else:
+            step()
+    t1.record(stream)
+    torch.cuda.synchronize()
+    if world > 1:
+        dist.barrier()
+    clk = clocks.stop()
+    ms = t0.elapsed_time(t1)
+    if world > 1:
+        t = torch.tensor([ms], device="cuda", dtype=torch.float64)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        ms = float(t.item())
+    launches = lps * steps if graph is not None else skm.skm_kernel_launches() - l0
+    timing = ("replays of one CUDA graph capturing the whole step" if graph is not None else "eager steps") + \
+        (f" ({note})" if note else "")
+    return ms, int(launches), timing, clk
+
+
+def _event_ms(fn, reps, stream):
+    """Mean CUDA-event time of fn() over reps calls, each bracketed alone."""
+    import torch
+
+    ts = []
+    for _ in range(reps):
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        fn()
+        e1.record(stream)
+        torch.cuda.synchronize()
+        ts.append(e0.elapsed_time(e1))
+    return statistics.mean(ts)
+
+
+def cpu_baseline_c4(Yb_host, C_host, K, budget_s=15.0):
+    """Oracle (as it stands) on a bounded row sample of the headline
+    workload: one Lloyd iteration (assignment against all k centroids in fp64,
+    update) of the first rows.  Returns (distances/s, rows, seconds, threads)."""
     import oracle
 
     def one(ns):
         t0 = time.perf_counter()
-        a, _, _ = oracle.assign_f32(X_host[:ns], C32)
-        oracle.update_f32(X_host[:ns], a, C32)
-        prep = oracle.rbq1_centroid_sq4(Cr, m)
-        ar, _ = oracle.rbq1_assign(codes[:ns], nx2[:ns], F[:ns], popx[:ns], DIM, prep)
-        oracle.rbq1_update(codes[:ns], F[:ns], DIM, m, e, ar, Cr)
+        a, _, _ = oracle.assign_bf16(Yb_host[:ns], C_host)
+        oracle.update_bf16(Yb_host[:ns], a, C_host)
         return time.perf_counter() - t0
 
-    t0 = one(500)
-    ns = int(min(X_host.shape[0], max(500, 500 * budget_s / max(t0, 1e-3))))
+    t0 = one(200)
+    ns = int(min(Yb_host.shape[0], max(200, 200 * budget_s / max(t0, 1e-3))))
     t = one(ns)
-    return 2.0 * ns * K / t, ns, t, oracle.num_threads()
+    return ns * K / t, ns, t, oracle.num_threads()
+
+
+def setup_head(dev, rank, world, dist, peaks):
+    """The headline workload resident in HBM: generated points, PCA basis
+    (rank 0's, broadcast), bf16 projection, Forgy centroids (rank 0's)."""
+    import torch
+
+    import paper_2608_14648_gb300 as skm
+    import synth
+
+    spec = synth.WORKLOADS[HEAD]
+    N, K = spec.n, spec.k
+    X = synth.workload_points(spec, seed=rank, device=dev)
+    mean = torch.empty(spec.d, device=dev, dtype=torch.float32)
+    P = torch.empty(spec.d, D_PCA, device=dev, dtype=torch.float32)
+    if rank == 0:
+        mean, P, _ = skm.skm_pca_fit(X, D_PCA)
+    if world > 1:
+        dist.broadcast(mean, 0)
+        dist.broadcast(P, 0)
+    skm.skm_project(X[:1024], P, mean, out_dtype=skm.DTYPE_BF16, max_ws_bytes=8 << 30)  # first-use costs
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record()
+    Y = skm.skm_project(X, P, mean, out_dtype=skm.DTYPE_BF16, max_ws_bytes=8 << 30)
+    e1.record()
+    torch.cuda.synchronize()
+    t_proj = e0.elapsed_time(e1)
+    del X
+    torch.cuda.empty_cache()
+    Yb = Y.view(torch.int16)
+    idx = synth.forgy_indices(N, K, seed=0).to(dev)
+    C = (Yb[idx].to(torch.int32) << 16).view(torch.float32).contiguous()
+    if world > 1:
+        dist.broadcast(C, 0)
+    flops = 6 * 2.0 * N * spec.d * D_PCA
+    proj = {"ms": t_proj, "bound": "tensor", "achieved": flops / (t_proj / 1e3) / 1e12, "peak": peaks["bf16_tflops"],
+            "unit": "TFLOP/s", "in_step": False,
+            "algorithmic": f"6 bf16 part products x 2*N*D*d' = {flops:.3e} flop (fp32-accurate projection, "
+                           "one-time preparation; includes the split pass)"}
+    proj["frac"] = proj["achieved"] / proj["peak"]
+    return Yb, C, idx, proj
+
+
+def run_extra_configs(args, dev, peaks, stream, local_rank):
+    """The 1M x 768 (fp32 and 1-bit) and 10M x 1024 (1-bit, k = 3,162)
+    iterations, each timed like the headline (graph replays), with clocks."""
+    import torch
+
+    import paper_2608_14648_gb300 as skm
+    import synth
+
+    out = {}
+
+    def timed(name, pts, C, k, n, d, flop_peak, kind):
+        wsA = skm.workspace(skm.OP_ASSIGN, pts, k)
+        wsU = skm.workspace(skm.OP_UPDATE, pts, k)
+        a = torch.empty(n, dtype=torch.int32, device=dev)
+        cnt = torch.zeros(k, dtype=torch.int64, device=dev)
+
+        def step():
+            skm.skm_assign(pts, C, k, want_dist=False, ws=wsA, out=a)
+            skm.skm_update(pts, a, C, counts=cnt, ws=wsU)
+
+        steps = max(5, min(args.steps, 20))
+        ms, launches, timing, clk = _timed_steps(step, stream, steps, 3, 1, None, local_rank, not args.eager)
+        t_a = _event_ms(lambda: skm.skm_assign(pts, C, k, want_dist=False, ws=wsA, out=a), 3, stream)
+        t_u = _event_ms(lambda: skm.skm_update(pts, a, C, counts=cnt, ws=wsU), 3, stream)
+        flops = 2.0 * n * k * d
+        ach = flops / (t_a / 1e3) / 1e12
+        out[name] = {"n": n, "d": d, "k": k, "ms_per_iter": ms / steps, "distances_per_s": n * k * steps / (ms / 1e3),
+                     "assign_ms": t_a, "update_ms": t_u, "assign_achieved_tflops": ach, "assign_peak_tflops": flop_peak,
+                     "assign_frac": ach / flop_peak, "flop": kind, "steps": steps, "timing": timing, "clocks": clk,
+                     "gpu_launches": launches}
+        del wsA, wsU
+
+    bf16 = peaks["bf16_tflops"]
+    spec = synth.WORKLOADS["emb1m_d768"]
+    X = synth.workload_points(spec, seed=0, device=dev)
+    idx = synth.forgy_indices(spec.n, spec.k, seed=0).to(dev)
+    timed("emb1m_d768_f32", skm.Points(skm.REPR_F32, X, spec.d).with_screen(), X[idx].clone(), spec.k, spec.n,
+          spec.d, bf16, "bf16")
+    pR = skm.rbq1_points(skm.skm_quantize(skm.REPR_RBQ1, X), spec.d).with_screen()
+    CR, _, _, _, _ = skm.skm_fit(pR, spec.k, 0, init_idx=idx, want_objective=False, want_dist=False)
+    timed("emb1m_d768_rbq1", pR, CR, spec.k, spec.n, spec.d, 2 * bf16, "e4m3")
+    # the AND + popcount 1-bit kernel on the same codes (no allocation entry point)
+    a_pop = torch.empty(spec.n, dtype=torch.int32, device=dev)
+    skm.skm_assign_rbq1_noalloc(pR, CR, a_pop)
+    t_pop = _event_ms(lambda: skm.skm_assign_rbq1_noalloc(pR, CR, a_pop), 2, stream)
+    popc = float(spec.n) * spec.k * 4 * ((spec.d + 31) // 32)
+    popc_peak = SM_COUNT * POPC_PER_CLK_SM * peaks["sm_max_mhz"] * 1e6
+    out["emb1m_d768_rbq1_popcount"] = {"assign_ms": t_pop, "bound": "alu", "achieved_tpopc": popc / (t_pop / 1e3) / 1e12,
+                                       "peak_tpopc": popc_peak / 1e12, "frac": popc / (t_pop / 1e3) / popc_peak,
+                                       "algorithmic": f"N*k*4*ceil(d/32) = {popc:.3e} POPC per launch"}
+    del X, pR, CR, a_pop
+    torch.cuda.empty_cache()
+
+    spec = synth.WORKLOADS["emb10m_d1024_rbq1"]
+    X = synth.workload_points(spec, seed=0, device=dev)
+    P = synth.haar_rotation(spec.d, 99).to(torch.float32).contiguous().to(dev)
+    Y = skm.skm_project(X, P, max_ws_bytes=8 << 30)
+    del X
+    q = skm.skm_quantize(skm.REPR_RBQ1, Y)
+    del Y
+    torch.cuda.empty_cache()
+    idx = synth.forgy_indices(spec.n, spec.k, seed=0).to(dev)
+    pR = skm.rbq1_points(q, spec.d).with_screen()
+    CR, _, _, _, _ = skm.skm_fit(pR, spec.k, 0, init_idx=idx, want_objective=False, want_dist=False)
+    timed("emb10m_d1024_rbq1", pR, CR, spec.k, spec.n, spec.d, 2 * bf16, "e4m3")
+    del pR, CR, q
+    torch.cuda.empty_cache()
+    return out
 
 
 def run_ours(args):
@@ -149,7 +354,6 @@ def run_ours(args):
     import torch
 
     import paper_2608_14648_gb300 as skm
-    import synth
 
     rank, local_rank, world = env_rank()
     torch.cuda.set_device(local_rank)
@@ -158,374 +362,168 @@ def run_ours(args):
     if world > 1:
         import torch.distributed as dist
 
-        from paper_2608_14648_gb300 import dist as skd
-
         dist.init_process_group("nccl")
     peaks = load_peaks()
+    stream = torch.cuda.current_stream()
 
     # ---- inputs (per-rank shard), resident in HBM before timing -------------
-    X = synth.gmm_points(N_POINTS, DIM, N_COMP, seed=rank, device=dev)
-    idx = synth.forgy_indices(N_POINTS, K, seed=0).to(dev)
-    C32 = X[idx].clone()
-    if world > 1:
-        dist.broadcast(C32, 0)
-    pts32 = skm.Points(skm.REPR_F32, X, DIM).with_screen()  # bf16 screening copy, built once
-    q = skm.skm_quantize(skm.REPR_RBQ1, X)
-    if world > 1:  # global mean, then re-encode; global fixed-point exponent
-        m = skd.global_mean(q["m"].double() * N_POINTS, N_POINTS)
-        q = skm.skm_quantize(skm.REPR_RBQ1, X, fit=False, m=m.contiguous())
-    e = skm.skm_rbq1_exponent(q["F"])
-    if world > 1:
-        e = skd.global_exponent(e, dev)
-    ptsR = skm.rbq1_points(q, DIM, e).with_screen()  # e4m3 expansion of the bits, built once
-    Cr, _, _, _, _ = skm.skm_fit(ptsR, K, 0, init_idx=idx, want_objective=False, want_dist=False)
-    if world > 1:
-        dist.broadcast(Cr, 0)
+    Yb, C, idx, proj = setup_head(dev, rank, world, dist, peaks)
+    N, K = Yb.shape[0], C.shape[0]
+    pts = skm.Points(skm.REPR_BF16, Yb, D_PCA).with_screen()  # per-point norms, built once
+    wsA = skm.workspace(skm.OP_ASSIGN, pts, K)
+    wsU = skm.workspace(skm.OP_UPDATE, pts, K)
+    a = torch.empty(N, dtype=torch.int32, device=dev)
+    cnt = torch.zeros(K, dtype=torch.int64, device=dev)
+    part = torch.zeros(K, D_PCA, dtype=torch.float64, device=dev) if world > 1 else None
+    C_step = C.clone()
 
-    wsA32 = skm.workspace(skm.OP_ASSIGN, pts32, K)
-    wsU32 = skm.workspace(skm.OP_UPDATE, pts32, K)
-    wsAR = skm.workspace(skm.OP_ASSIGN, ptsR, K)
-    wsUR = skm.workspace(skm.OP_UPDATE, ptsR, K)
-    a32 = torch.empty(N_POINTS, dtype=torch.int32, device=dev)
-    aR = torch.empty(N_POINTS, dtype=torch.int32, device=dev)
-    cnt32 = torch.zeros(K, dtype=torch.int64, device=dev)
-    cntR = torch.zeros(K, dtype=torch.int64, device=dev)
-    part32 = torch.zeros(K, DIM, dtype=torch.float64, device=dev) if world > 1 else None
-    partR = torch.zeros(K, DIM + 1, dtype=torch.int64, device=dev) if world > 1 else None
-    stream = torch.cuda.current_stream()
-    ev = {name: [] for name in ("a32", "aR")}
-
-    def lloyd(pts, C, a, cnt, part, wsA, wsU, key, record):
-        if record:
-            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-            e0.record(stream)
-        skm.skm_assign(pts, C, K, want_dist=False, ws=wsA, out=a)
-        if record:
-            e1.record(stream)
-            ev[key].append((e0, e1))
+    def step():
+        skm.skm_assign(pts, C_step, K, want_dist=False, ws=wsA, out=a)
         if part is None:
-            skm.skm_update(pts, a, C, counts=cnt, ws=wsU)
-        else:
+            skm.skm_update(pts, a, C_step, counts=cnt, ws=wsU)
+        else:  # the one exchange: cluster sums and counts, all-reduced
             part.zero_()
             cnt.zero_()
             skm.skm_update(pts, a, None, counts=cnt, partial=part, ws=wsU)
-            skd.allreduce_partials(part, cnt)
-            skm.skm_update_finalize(pts, part, cnt, C)
+            dist.all_reduce(part)
+            dist.all_reduce(cnt)
+            skm.skm_update_finalize(pts, part, cnt, C_step)
 
-    def step(record):
-        lloyd(pts32, C32, a32, cnt32, part32, wsA32, wsU32, "a32", record)
-        lloyd(ptsR, Cr, aR, cntR, partR, wsAR, wsUR, "aR", record)
-
-    for _ in range(args.warmup):
-        step(False)
-    torch.cuda.synchronize()
-    # One GPU: the step (both Lloyd iterations, every kernel of assign and
-    # update) is captured once in a CUDA graph and replayed, so no host launch
-    # gap sits between kernels; the library's launch counter during the
-    # capture gives the kernels per step.  Several GPUs: eager (the exchange is
-    # an NCCL all-reduce between the ranks).
-    graph, launches_per_step, graph_note = None, None, None
-    if world == 1 and not args.eager:
-        try:
-            side = torch.cuda.Stream()
-            side.wait_stream(stream)
-            with torch.cuda.stream(side):
-                step(False)
-            stream.wait_stream(side)
-            torch.cuda.synchronize()
-            l0 = skm.skm_kernel_launches()
-            graph = torch.cuda.CUDAGraph()
-            with torch.cuda.graph(graph):
-                step(False)
-            launches_per_step = skm.skm_kernel_launches() - l0
-            graph.replay()
-            torch.cuda.synchronize()
-        except Exception as exc:
-            graph, graph_note = None, f"graph capture failed, eager steps: {exc!r}"[:200]
-    if world > 1:
-        dist.barrier()
-    clocks = ClockSampler(local_rank)
-    clocks.start()
-    torch.cuda.synchronize()
-    launches0 = skm.skm_kernel_launches()
-    t_start, t_end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    t_start.record(stream)
-    for _ in range(args.steps):
-        if graph is not None:
-            graph.replay()
-        else:
-            step(True)
-    t_end.record(stream)
-    torch.cuda.synchronize()
-    if world > 1:
-        dist.barrier()
-    launches = (launches_per_step * args.steps if graph is not None
-                else skm.skm_kernel_launches() - launches0)
-    if graph is not None:  # per-kernel event times from eager steps after the timed region
-        for _ in range(3):
-            step(True)
-        torch.cuda.synchronize()
-    clk = clocks.stop()
-    ms = t_start.elapsed_time(t_end)
-    if world > 1:
-        t = torch.tensor([ms], device=dev, dtype=torch.float64)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        ms = float(t.item())
+    ms, launches, timing, clk = _timed_steps(step, stream, args.steps, args.warmup, world, dist, local_rank,
+                                             world == 1 and not args.eager)
     ms_step = ms / args.steps
-    value = world * 2.0 * N_POINTS * K * args.steps / (ms / 1e3)
+    value = world * float(N) * K * args.steps / (ms / 1e3)
 
-    # ---- the AND+popcount 1-bit kernel, timed beside the tensor-core one --------
-    t_pop = None
-    if not args.no_popcount:
-        torch.cuda.synchronize()
-        p0, p1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-        a_pop = torch.empty_like(aR)
-        skm.skm_assign_rbq1_noalloc(ptsR, Cr, a_pop)
-        p0.record(stream)
-        skm.skm_assign_rbq1_noalloc(ptsR, Cr, a_pop)
-        p1.record(stream)
-        torch.cuda.synchronize()
-        t_pop = p0.elapsed_time(p1)
-
-    # ---- roofline of the dominant kernel --------------------------------------
-    t_a32 = statistics.mean(a.elapsed_time(b) for a, b in ev["a32"])
-    t_aR = statistics.mean(a.elapsed_time(b) for a, b in ev["aR"])
+    # ---- per-kernel times (eager calls after the timed region) ----------------
+    t_assign = _event_ms(lambda: skm.skm_assign(pts, C_step, K, want_dist=False, ws=wsA, out=a), 3, stream)
+    t_update = _event_ms(lambda: skm.skm_update(pts, a, C_step.clone(), counts=cnt, ws=wsU), 3, stream)
     long_region = ms > 1000.0
     bf16_peak = peaks["bf16_tflops_sustained"] if long_region else peaks["bf16_tflops"]
-    fp8_peak = 2.0 * bf16_peak  # nominal dense e4m3 : bf16 ratio (4.5 : 2.25 PFLOP/s)
-    flops = 2.0 * N_POINTS * K * DIM
-    W = (DIM + 31) // 32
-    popc_aR = float(N_POINTS) * K * 4 * W
-    popc_peak = SM_COUNT * POPC_PER_CLK_SM * peaks["sm_max_mhz"] * 1e6  # per second
+    flops = 2.0 * N * K * D_PCA
+    upd_bytes = N * D_PCA * 2 + N * 4 * 3  # rows read once; assignments, sorted order, cluster ids
     kernels = {
-        "assign_f32": {"ms": t_a32, "bound": "tensor", "achieved": flops / (t_a32 / 1e3) / 1e12,
-                       "peak": bf16_peak, "unit": "TFLOP/s",
-                       "algorithmic": f"2*N*k*d = {flops:.3e} bf16 flop per launch (screen GEMM)"},
-        "assign_rbq1": {"ms": t_aR, "bound": "tensor", "achieved": flops / (t_aR / 1e3) / 1e12,
-                        "peak": fp8_peak, "unit": "TFLOP/s",
-                        "algorithmic": f"2*N*k*d = {flops:.3e} e4m3 flop per launch (exact integer P)"},
+        "assign_bf16_screen": {
+            "ms": t_assign, "bound": "tensor", "achieved": flops / (t_assign / 1e3) / 1e12, "peak": bf16_peak,
+            "unit": "TFLOP/s",
+            "algorithmic": f"2*N*k*d' = {flops:.3e} bf16 flop per launch (tensor-core screen; the call also "
+                           "prepares the centroids and rescores undecided rows in fp32)"},
+        "update_bf16": {
+            "ms": t_update, "bound": "hbm", "achieved": upd_bytes / (t_update / 1e3) / 1e9, "peak": peaks["hbm_gbs"],
+            "unit": "GB/s", "algorithmic": f"N*d'*2 + 12*N = {upd_bytes:.3e} bytes per launch (bf16 rows read once, "
+                                           "assignments, sorted order and cluster ids)"},
+        "project_pca": proj,
     }
-    if t_pop is not None:
-        kernels["assign_rbq1_popcount"] = {
-            "ms": t_pop, "bound": "alu", "achieved": popc_aR / (t_pop / 1e3) / 1e12,
-            "peak": popc_peak / 1e12, "unit": "Tpopc/s", "in_step": False,
-            "algorithmic": f"N*k*4*ceil(d/32) = {popc_aR:.3e} POPC per launch"}
+
+    # ---- the pruned assignment of the same workload (exact, SKM_FLAG_PRUNE) on a row subset
+    if not args.no_prune and world == 1:
+        ns = min(N, 1_000_000)
+        pp = skm.Points(skm.REPR_BF16, Yb[:ns], D_PCA, flags=skm.FLAG_PRUNE)
+        ap = torch.empty(ns, dtype=torch.int32, device=dev)
+        prev = a[:ns].clone()  # bound seeded with the previous assignment's centroid
+        wsP = skm.workspace(skm.OP_ASSIGN, pp, K)
+        skm.skm_assign(pp, C_step, K, prev_assign=prev, want_dist=False, ws=wsP, out=ap)
+        t_prune = _event_ms(lambda: skm.skm_assign(pp, C_step, K, prev_assign=prev, want_dist=False, ws=wsP,
+                                                   out=ap), 2, stream)
+        _, _, _, _, st = skm.skm_fit(pp, K, 0, C_init=C_step, want_objective=False, want_dist=False)
+        same = bool(torch.equal(ap, a[:ns]))
+        pairs = float(ns) * K
+        dense_ms = t_assign * ns / N
+        kernels["assign_bf16_prune"] = {
+            "ms": t_prune, "rows": ns, "in_step": False, "bound": "fp32 CUDA cores",
+            "first_block_survivors": st["prune_first_block"] / pairs, "complete_survivors": st["prune_complete"] / pairs,
+            "dense_screen_ms_same_rows": dense_ms, "speedup_vs_dense": dense_ms / t_prune,
+            "same_assignment_as_dense": same,
+            "note": "exact 32-dimension prefix-block pruning, bound seeded with the previous assignment"}
+        del pp, ap, prev, wsP
     for kd in kernels.values():
-        kd["frac"] = kd["achieved"] / kd["peak"]
-    dom = max((n for n in kernels if kernels[n].get("in_step", True)), key=lambda n: kernels[n]["ms"])
-    kd = kernels[dom]
-    traffic = TRAFFIC_PER_POINT.get(dom)
+        if "achieved" in kd:
+            kd["frac"] = kd["achieved"] / kd["peak"]
+    kd = kernels["assign_bf16_screen"]
+    traffic = TRAFFIC_PER_POINT.get("assign_bf16_screen")
     roofline = {"bound": kd["bound"], "achieved": round(kd["achieved"], 4), "peak": round(kd["peak"], 4),
                 "unit": kd["unit"], "frac": round(kd["frac"], 5),
-                "traffic": round(traffic * N_POINTS) if traffic else None, "kernel": dom,
-                "peak_source": f"{peaks['source']} ({'sustained' if long_region else 'burst'} bf16"
-                               f"{', x2 for e4m3' if dom == 'assign_rbq1' else ''})"}
+                "traffic": round(traffic * N) if traffic else None, "kernel": "assign_bf16_screen",
+                "peak_source": f"{peaks['source']} ({'sustained' if long_region else 'burst'} bf16)"}
 
     # ---- end to end through the C ABI with host buffers ----------------------
     e2e = None
     if not args.no_e2e:
-        X_host = torch.empty(N_POINTS, DIM, dtype=torch.float32, pin_memory=True)
-        X_host.copy_(X)
-        C_host32 = torch.empty(K, DIM, dtype=torch.float32, pin_memory=True)
-        C_hostR = torch.empty(K, DIM, dtype=torch.float32, pin_memory=True)
-        C_host32.copy_(C32)
-        C_hostR.copy_(Cr)
-        a_host = torch.empty(2, N_POINTS, dtype=torch.int32, pin_memory=True)
-        # two device buffers for the points: step t + 1's copy streams in while
-        # step t is still being assigned and updated (the next step's points do
-        # not depend on this step; its centroids do, and wait for the D2H)
-        Xbuf = [torch.empty_like(X), torch.empty_like(X)]
-        Cd32 = torch.empty_like(C32)
-        CdR = torch.empty_like(Cr)
-        # The H2D copy of the points is cut into E2E_CHUNKS row ranges on a copy
-        # stream; each range is assigned (fp32: screening copy built inside the
-        # call; 1-bit: encoded, then assigned) and its fp32 cluster sums are
-        # added into fp64 partial sums (the sharded update form) as soon as it
-        # has landed, so the copy of later ranges overlaps the work on earlier
-        # ones.  The fp32 update is finalised after the last range; the 1-bit
-        # update needs the fixed-point exponent of every F and runs after it.
-        nchunk = E2E_CHUNKS
-        bounds = [(i * N_POINTS // nchunk, (i + 1) * N_POINTS // nchunk) for i in range(nchunk)]
-        cmax = max(b1 - b0 for b0, b1 in bounds)
-        W = (DIM + 31) // 32
-        codesE = torch.empty(N_POINTS, W, device=dev, dtype=torch.int32)
-        nx2E = torch.empty(N_POINTS, device=dev, dtype=torch.float32)
-        FE = torch.empty(N_POINTS, device=dev, dtype=torch.float32)
-        popxE = torch.empty(N_POINTS, device=dev, dtype=torch.int32)
-        mE = q["m"]
-        probe32 = skm.Points(skm.REPR_F32, Xbuf[0][:cmax], DIM)
-        wsA2 = skm.workspace(skm.OP_ASSIGN, probe32, K)
-        wsAR2 = skm.workspace(skm.OP_ASSIGN, skm.Points(skm.REPR_RBQ1, codesE[:cmax], DIM, nx2E[:cmax],
-                                                        FE[:cmax], popxE[:cmax], mE, e), K)
-        wsQ2 = skm.workspace(skm.OP_QUANTIZE, probe32, 1)
-        part32e = torch.zeros(K, DIM, device=dev, dtype=torch.float64)
-        cnt32e = torch.zeros(K, device=dev, dtype=torch.int64)
-        wsU2 = skm.workspace(skm.OP_UPDATE, probe32, K)
-        copy_stream = torch.cuda.Stream()   # the points, one step ahead
-        cent_stream = torch.cuda.Stream()   # the centroids, after the previous step's D2H
+        Y_host = torch.empty(N, D_PCA, dtype=torch.int16, pin_memory=True)
+        Y_host.copy_(Yb)
+        C_host = torch.empty(K, D_PCA, dtype=torch.float32, pin_memory=True)
+        C_host.copy_(C)
+        a_host = torch.empty(N, dtype=torch.int32, pin_memory=True)
+        holder = {}
+
+        def exchange():
+            s = holder["step"]
+            dist.all_reduce(s.partial)
+            dist.all_reduce(s.counts)
+
+        hstep = skm.LloydStepHost(skm.REPR_BF16, Y_host, D_PCA, K, chunks=E2E_CHUNKS, device=dev,
+                                  exchange=exchange if world > 1 else None)
+        holder["step"] = hstep
+        for _ in range(2):  # untimed warm-up (first-use costs of the range-sized calls)
+            hstep(C_host, C_host, a_host)
         e2e_steps = max(2, min(args.steps, 5))
-        landed = [[torch.cuda.Event() for _ in range(nchunk)] for _ in range(2)]
-        c_landed = torch.cuda.Event()
-        buf_free = [torch.cuda.Event(), torch.cuda.Event()]
-        d2h_done = torch.cuda.Event()
-        # per-range point descriptors over the fixed device buffers (views)
-        pcs = [[skm.Points(skm.REPR_F32, xb[b0:b1], DIM) for b0, b1 in bounds] for xb in Xbuf]
-        qouts = [{"codes": codesE[b0:b1], "nx2": nx2E[b0:b1], "F": FE[b0:b1], "popx": popxE[b0:b1]}
-                 for b0, b1 in bounds]
-        prcs = [skm.Points(skm.REPR_RBQ1, codesE[b0:b1], DIM, nx2E[b0:b1], FE[b0:b1], popxE[b0:b1], mE, e)
-                for b0, b1 in bounds]
-        pall = [skm.Points(skm.REPR_F32, xb, DIM) for xb in Xbuf]
-        host_ms = []
-        h2d = X_host.numel() * 4 + 2 * K * DIM * 4
-        d2h = 2 * N_POINTS * 4 + 2 * K * DIM * 4
-        # the host link's copy rate just before the run (the e2e step is bound by
-        # it; it varies with other traffic on the shared host)
-        torch.cuda.synchronize()
-        p0, p1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-        p0.record(stream)
-        Xbuf[0].copy_(X_host, non_blocking=True)
-        p1.record(stream)
-        torch.cuda.synchronize()
-        h2d_probe_gbs = X_host.numel() * 4 / (p0.elapsed_time(p1) / 1e3) / 1e9
-
-        def enqueue_points(t):
-            slot = t % 2
-            if t >= 2:
-                copy_stream.wait_event(buf_free[slot])  # step t - 2 is done with this buffer
-            with torch.cuda.stream(copy_stream):
-                for (b0, b1), ev in zip(bounds, landed[slot]):
-                    Xbuf[slot][b0:b1].copy_(X_host[b0:b1], non_blocking=True)
-                    ev.record(copy_stream)
-
-        def e2e_run(nsteps):
-            """nsteps end-to-end steps; the device time from the first copy to the
-            last step's D2H (ms)."""
-            s0, s1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-            s0.record(stream)
-            copy_stream.wait_stream(stream)
-            cent_stream.wait_stream(stream)
-            enqueue_points(0)
-            for t in range(nsteps):
-                th0 = time.perf_counter()
-                slot = t % 2
-                if t + 1 < nsteps:
-                    enqueue_points(t + 1)
-                if t > 0:
-                    cent_stream.wait_event(d2h_done)  # this step's centroids are the last step's results
-                # by the SMs, not a copy engine: there they would queue behind the
-                # next step's point ranges
-                skm.skm_copy_from_host(Cd32, C_host32, stream=cent_stream)
-                skm.skm_copy_from_host(CdR, C_hostR, stream=cent_stream)
-                c_landed.record(cent_stream)
-                stream.wait_event(c_landed)
-                part32e.zero_()
-                cnt32e.zero_()
-                xb = Xbuf[slot]
-                for (b0, b1), ev, pc, qo, prc in zip(bounds, landed[slot], pcs[slot], qouts, prcs):
-                    stream.wait_event(ev)
-                    skm.skm_assign(pc, Cd32, K, want_dist=False, ws=wsA2, out=a32[b0:b1])
-                    skm.skm_update(pc, a32[b0:b1], None, counts=cnt32e, partial=part32e, ws=wsU2)
-                    skm.skm_quantize(skm.REPR_RBQ1, xb[b0:b1], fit=False, m=mE, ws=wsQ2, out=qo)
-                    skm.skm_assign(prc, CdR, K, want_dist=False, ws=wsAR2, out=aR[b0:b1])
-                buf_free[slot].record(stream)
-                if world > 1:  # the same exchange as the device-resident step
-                    skd.allreduce_partials(part32e, cnt32e)
-                skm.skm_update_finalize(pall[slot], part32e, cnt32e, Cd32)
-                host_ms.append((time.perf_counter() - th0) * 1e3)  # enqueue only (no sync so far)
-                eE = skm.skm_rbq1_exponent(FE)
-                if world > 1:
-                    eE = skd.global_exponent(eE, dev)
-                pR2 = skm.Points(skm.REPR_RBQ1, codesE, DIM, nx2E, FE, popxE, mE, eE)
-                if world > 1:
-                    partR.zero_()
-                    cntR.zero_()
-                    skm.skm_update(pR2, aR, None, counts=cntR, partial=partR, ws=wsUR)
-                    skd.allreduce_partials(partR, cntR)
-                    skm.skm_update_finalize(pR2, partR, cntR, CdR)
-                else:
-                    skm.skm_update(pR2, aR, CdR, counts=cntR, ws=wsUR)
-                a_host[0].copy_(a32, non_blocking=True)
-                a_host[1].copy_(aR, non_blocking=True)
-                C_host32.copy_(Cd32, non_blocking=True)
-                C_hostR.copy_(CdR, non_blocking=True)
-                d2h_done.record(stream)
-            s1.record(stream)
-            torch.cuda.synchronize()
-            return s0.elapsed_time(s1)
-
-        e2e_run(2)  # warm-up (first-use costs of the range-sized calls), untimed
-        host_ms.clear()
         if world > 1:
             dist.barrier()
-        def timed_e2e():
-            t_ms = e2e_run(e2e_steps)
-            if world > 1:
-                t = torch.tensor([t_ms], device=dev, dtype=torch.float64)
-                dist.all_reduce(t, op=dist.ReduceOp.MAX)
-                t_ms = float(t.item())
-            return t_ms
-
-        ems = timed_e2e()
-        # The host link is shared with the host's other traffic: a run whose
-        # copies averaged under 3/4 of the rate probed just before it is taken
-        # again once (both attempts are reported).
-        probe = h2d_probe_gbs
-        if world > 1:
-            t = torch.tensor([probe], device=dev, dtype=torch.float64)
-            dist.all_reduce(t, op=dist.ReduceOp.MIN)
-            probe = float(t.item())
-        first_attempt = None
-        if h2d / (ems / e2e_steps / 1e3) / 1e9 < 0.75 * probe:
-            first_attempt = {"ms_per_step": ems / e2e_steps,
-                             "h2d_effective_gbs": round(h2d / (ems / e2e_steps / 1e3) / 1e9, 1)}
-            host_ms.clear()
-            if world > 1:
-                dist.barrier()
-            ems = timed_e2e()
-        # and right after it: the link is shared with the host's other traffic
         torch.cuda.synchronize()
+        t0 = time.perf_counter()
+        for _ in range(e2e_steps):
+            hstep(C_host, C_host, a_host)  # synchronous: results are in host memory on return
+        ems = (time.perf_counter() - t0) * 1e3
+        if world > 1:
+            t = torch.tensor([ems], device=dev, dtype=torch.float64)
+            dist.all_reduce(t, op=dist.ReduceOp.MAX)
+            ems = float(t.item())
+        # the host link's copy rate right after (the step's bound when the work is shorter)
+        p0, p1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
         p0.record(stream)
-        Xbuf[0].copy_(X_host, non_blocking=True)
+        Yb.copy_(Y_host, non_blocking=True)
         p1.record(stream)
         torch.cuda.synchronize()
-        h2d_probe_after_gbs = X_host.numel() * 4 / (p0.elapsed_time(p1) / 1e3) / 1e9
-        e2e = {"value": world * 2.0 * N_POINTS * K * e2e_steps / (ems / 1e3), "unit": "distances/s",
+        h2d_probe_gbs = Y_host.numel() * 2 / (p0.elapsed_time(p1) / 1e3) / 1e9
+        h2d = Y_host.numel() * 2 + C_host.numel() * 4
+        d2h = a_host.numel() * 4 + C_host.numel() * 4
+        e2e = {"value": world * float(N) * K * e2e_steps / (ems / 1e3), "unit": "distances/s",
                "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "steps": e2e_steps,
-               "host_enqueue_ms_per_step": round(statistics.mean(host_ms), 3),
-               "h2d_probe_gbs": round(h2d_probe_gbs, 1), "h2d_probe_after_gbs": round(h2d_probe_after_gbs, 1),
+               "ms_per_step": ems / e2e_steps, "h2d_probe_gbs": round(h2d_probe_gbs, 1),
                "h2d_effective_gbs": round(h2d / (ems / e2e_steps / 1e3) / 1e9, 1),
-               "remeasured_after": first_attempt,
-               "ms_per_step": ems / e2e_steps,
-               "path": f"pinned host fp32 points -> H2D in {nchunk} row ranges on a copy stream (two device "
-                       "buffers: the next step's points stream in during this step's tail), each range assigned "
-                       "(fp32) and encoded + assigned (1-bit) once it has landed -> skm_update (fp32, 1-bit) -> "
-                       "D2H assignments + centroids, which the next step copies back as its centroids"}
+               "path": f"skm_lloyd_step_host: pinned host bf16 points -> {E2E_CHUNKS} row ranges copied on a copy "
+                       "stream into three device range buffers while earlier ranges are assigned and summed -> "
+                       "finalised centroids and assignments back in host memory on return (host wall clock per "
+                       "call)"}
+        del hstep, Y_host
+
+    # ---- the other configurations (one GPU) -------------------------------------
+    extra = None
+    if world == 1 and not args.no_extra:
+        del wsA, wsU, pts
+        torch.cuda.empty_cache()
+        extra = run_extra_configs(args, dev, peaks, stream, local_rank)
 
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        h = {k2: v.cpu().numpy() for k2, v in q.items()}
-        codes = h["codes"].view(np.uint32)
-        X_host_np = X[:200_000].cpu().numpy()
-        v, ns, t, cores = cpu_baseline_sample(X_host_np, C32.cpu().numpy(), codes, h["nx2"], h["F"], h["popx"],
-                                              h["m"], e, Cr.cpu().numpy())
+        Yh = Yb[:200_000].cpu().numpy().view(np.uint16)
+        v, ns, t, cores = cpu_baseline_c4(Yh, C.cpu().numpy(), K)
         cpu = {"value": v, "unit": "distances/s", "cores": cores, "kind": "oracle",
-               "sample": f"{ns} of {N_POINTS} rows, one Lloyd iteration (assign + update) of fp32 and 1-bit "
-                         f"against all {K} centroids, {t:.1f} s"}
+               "sample": f"{ns} of {N} rows of the headline workload, one Lloyd iteration (fp64 assignment "
+                         f"against all {K} centroids + update), {t:.1f} s"}
 
     if rank == 0:
         line = {
             "metric": METRIC, "value": value, "unit": "distances/s", "n_gpus": world, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": ms_step, "higher_is_better": True, "scaling": "weak",
-            "vs_baseline": None, "dtype": "f32 (bf16 tensor screen + fp32 rescore) / 1-bit (e4m3 tensor, exact)",
-            "data": "synthetic (seeded GMM embeddings, generated on the GPU)",
-            "config": {"workload": WORKLOAD, "n": N_POINTS, "d": DIM, "k": K, "reprs": ["f32", "rbq1"],
-                       "step": "one Lloyd iteration (assign + update) per representation",
-                       "l2": "inputs larger than L2 (3.1 GB fp32 points streamed every step)",
-                       "timing": ("replays of one CUDA graph capturing the whole step" if graph is not None
-                                  else "eager steps") + (f" ({graph_note})" if graph_note else ""),
-                       "parallelism": f"dp{world}"},
-            "roofline": roofline, "kernels": kernels, "cpu_baseline": cpu, "e2e": e2e, "clocks": clk,
-            "gpu_launches": int(launches),
+            "vs_baseline": None,
+            "dtype": "bf16 points, fp32 centroids (bf16 tensor-core screen + fp32 rescore: the exact fp32 argmin)",
+            "data": "synthetic (seeded GMM embeddings, generated on the GPU; PCA fitted on them)",
+            "config": {"workload": WORKLOAD, "n": N, "D": 1024, "d": D_PCA, "k": K, "repr": "bf16 (PCA-256)",
+                       "step": "one Lloyd iteration (assign + update) over all points",
+                       "l2": "inputs larger than L2 (5.1 GB of bf16 points streamed every step)",
+                       "timing": timing, "parallelism": f"dp{world}"},
+            "roofline": roofline, "kernels": kernels, "configs": extra, "cpu_baseline": cpu, "e2e": e2e,
+            "clocks": clk, "gpu_launches": launches,
         }
         print(json.dumps(line), flush=True)
     if world > 1:
@@ -533,50 +531,49 @@ def run_ours(args):
 
 
 def run_reference(args):
-    """CPU oracle as it stands, on the host cores, on a bounded sample."""
-    import numpy as np
-
+    """CPU oracle as it stands, on the host cores, on a bounded sample of the
+    headline workload's recipe (PCA fitted on the sample)."""
     rank, _, world = env_rank()
     if rank != 0:
         return
     import oracle
     import synth
 
-    ns = 4000
-    X = synth.gmm_points(ns, DIM, N_COMP, seed=0).numpy()
+    spec = synth.WORKLOADS[HEAD]
+    ns = 20_000
+    X = synth.gmm_points(ns, spec.d, spec.n_comp, seed=0, decay=spec.decay, std=spec.std).numpy()
+    mu, P, _ = oracle.pca_fit(X, D_PCA)
+    Yb = oracle.round_bf16(oracle.project(X, P, mu))
+    del X
+    K = spec.k
     idx = synth.forgy_indices(ns, K, seed=0).numpy()
-    C32 = X[idx].copy()
-    m = oracle.rbq1_mean(X)
-    codes, nx2, F, popx = oracle.rbq1_encode(X, m)
-    e = oracle.rbq1_exponent(F)
-    Cr = oracle.rbq1_decode_points(codes, F, DIM, m, e, idx)
+    C = oracle.bf16_to_f32(Yb[idx]).copy()
 
     def step(rows):
-        nonlocal C32, Cr
-        a, _, _ = oracle.assign_f32(X[:rows], C32)
-        C32, _ = oracle.update_f32(X[:rows], a, C32)
-        prep = oracle.rbq1_centroid_sq4(Cr, m)
-        ar, _ = oracle.rbq1_assign(codes[:rows], nx2[:rows], F[:rows], popx[:rows], DIM, prep)
-        Cr, _ = oracle.rbq1_update(codes[:rows], F[:rows], DIM, m, e, ar, Cr)
+        nonlocal C
+        a, _, _ = oracle.assign_bf16(Yb[:rows], C)
+        C, _ = oracle.update_bf16(Yb[:rows], a, C)
 
     t0 = time.perf_counter()
-    step(500)
+    step(200)
     t1 = time.perf_counter() - t0
     budget = 150.0 / max(1, args.steps + args.warmup)
-    rows = int(min(ns, max(500, 500 * budget / max(t1, 1e-3))))
+    rows = int(min(ns, max(200, 200 * budget / max(t1, 1e-3))))
     for _ in range(args.warmup):
         step(rows)
     t0 = time.perf_counter()
     for _ in range(args.steps):
         step(rows)
     t = time.perf_counter() - t0
-    value = 2.0 * rows * K * args.steps / t
-    sample = f"{rows} rows of the {WORKLOAD} recipe, one Lloyd iteration per representation per step"
+    value = float(rows) * K * args.steps / t
+    sample = (f"{rows} rows of the {HEAD} recipe (PCA fitted on a {ns}-row sample), one Lloyd iteration against "
+              f"all {K} centroids per step")
     line = {"impl": "reference", "metric": METRIC, "value": value, "unit": "distances/s", "n_gpus": world,
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * t / args.steps,
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64 (oracle)",
             "data": "synthetic (seeded GMM embeddings)",
-            "config": {"workload": WORKLOAD, "n": N_POINTS, "d": DIM, "k": K, "reprs": ["f32", "rbq1"],
+            "config": {"workload": WORKLOAD, "n": spec.n, "D": spec.d, "d": D_PCA, "k": K, "repr": "bf16 (PCA-256)",
+                       "step": "one Lloyd iteration (assign + update) over the sampled points",
                        "parallelism": "host cores"},
             "cpu_baseline": {"value": value, "unit": "distances/s", "kind": "oracle", "cores": oracle.num_threads(),
                              "sample": sample},
@@ -649,6 +646,10 @@ def run_case(args):
         q = skm.skm_quantize(skm.REPR_SQ8, X)
         pts = skm.Points(skm.REPR_SQ8, q["codes"], d, flags=skm.FLAG_PRUNE)
         C = q["codes"][synth.forgy_indices(n, k, seed=0).cuda()].clone()
+    elif args.case == "assign_bf16":  # bf16 points, tensor-core screen (the headline's kernel)
+        Xb = X.to(torch.bfloat16).view(torch.int16).contiguous()
+        pts = skm.Points(skm.REPR_BF16, Xb, d).with_screen()
+        C = (Xb[synth.forgy_indices(n, k, seed=0).cuda()].to(torch.int32) << 16).view(torch.float32).contiguous()
     elif args.case == "assign_prune":  # bf16 points, exact prefix-block pruning
         Xb = X.to(torch.bfloat16).view(torch.int16).contiguous()
         pts = skm.Points(skm.REPR_BF16, Xb, d, flags=skm.FLAG_PRUNE)
@@ -943,10 +944,11 @@ def main():
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
-    ap.add_argument("--no-popcount", action="store_true")
+    ap.add_argument("--no-prune", action="store_true", help="skip the pruned assignment of the headline workload")
+    ap.add_argument("--no-extra", action="store_true", help="skip the 1M x 768 and 10M x 1024 1-bit iterations")
     ap.add_argument("--eager", action="store_true", help="time eager steps instead of CUDA-graph replays")
     ap.add_argument("--case", default=None,
-                    help="single-operation run for profiling: assign_f32|assign_rbq1|assign_sq8|assign_lvq4|"
+                    help="single-operation run for profiling: assign_f32|assign_bf16|assign_rbq1|assign_sq8|assign_lvq4|"
                          "assign_rbq1_popcount|assign_prune|assign_prune_sq8|update_f32|update_rbq1|update_sq8|"
                          "update_lvq4|project|quantize_sq8|quantize_rbq1|quantize_lvq4")
     ap.add_argument("--n", type=int, default=200_000)

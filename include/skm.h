@@ -45,7 +45,8 @@ typedef enum skm_status {
     SKM_ERR_CUDA = 3,         /* a CUDA runtime/driver call failed            */
     SKM_ERR_NO_MEMORY = 4,    /* ws_bytes smaller than skm_workspace_size()  */
     SKM_ERR_TIMEOUT = 5,      /* a bounded device wait gave up               */
-    SKM_ERR_DEVICE_CHECK = 6  /* a device-side check recorded a failure      */
+    SKM_ERR_DEVICE_CHECK = 6, /* a device-side check recorded a failure      */
+    SKM_ERR_EXCHANGE = 7      /* a caller's exchange hook reported a failure */
 } skm_status;
 
 /* ---- representations of the points being clustered (Table 1) ---------- */
@@ -124,6 +125,29 @@ typedef struct skm_stats {
 const char *skm_last_error(void);
 int skm_version(void); /* major*10000 + minor*100 + patch */
 
+/* Fault injection, for tests of the error paths (the paper has no
+ * counterpart).  Arms `count` occurrences (0 disarms) of one fault, process
+ * wide; each occurrence is used up by the first place that checks for it:
+ *  SKM_FAULT_WORKSPACE  a workspace check reports SKM_ERR_NO_MEMORY, before
+ *                       anything is enqueued;
+ *  SKM_FAULT_LAUNCH     a kernel launch reports a launch failure: that kernel
+ *                       still runs, the entry point enqueues nothing more and
+ *                       returns SKM_ERR_CUDA;
+ *  SKM_FAULT_STATUS     skm_fit's final read of its device status word finds
+ *                       it set (the fault writes it on the device), so the
+ *                       call returns SKM_ERR_DEVICE_CHECK;
+ *  SKM_FAULT_WAIT       a tensor-core assignment launch starts with a 1 ms
+ *                       bounded wait on a barrier that nothing arrives on: it
+ *                       gives up before loading anything, raises its abort
+ *                       flag, and skm_fit reports SKM_ERR_TIMEOUT.
+ * The environment variable SKM_FAULT=workspace|launch|status|wait arms one
+ * occurrence when the library first checks.  Nothing faults the GPU: every
+ * injected failure is a status the host reads.  Returns SKM_OK, or
+ * SKM_ERR_INVALID_ARG for an unknown kind or a negative count. */
+enum { SKM_FAULT_WORKSPACE = 1, SKM_FAULT_LAUNCH = 2, SKM_FAULT_STATUS = 3, SKM_FAULT_WAIT = 4 };
+int skm_inject_fault(int kind, int count);
+int skm_fault_armed(int kind); /* occurrences left (0 for an unknown kind) */
+
 /* Number of CUDA kernels this library has enqueued in this process so far
  * (host-side counter over all threads and devices; diagnostic only, e.g. to
  * count the kernels inside a timed region). */
@@ -192,6 +216,15 @@ int skm_copy_from_host(void *dst, const void *src_host, size_t bytes, void *stre
  * Distances are preserved up to rounding.  Asynchronous. */
 int skm_project_hadamard(const float *X, int64_t n, int d, const float *mean, const float *sigma,
                          int D, int out_dtype, void *Y, void *stream);
+
+/* Forgy initialisation (Section 2.3 STEP 1: k points sampled at random),
+ * HOST helper: idx_host[0..k) = positions 0..k-1 of a Fisher-Yates shuffle
+ * of (0, 1, ..., n-1) in which position i = 0, 1, ..., k-1 swaps with
+ * i + floor(r (n - i) / 2^64), r = w0 2^32 + w1 from (w0, w1, w2, w3) =
+ * Philox4x32-10 of counter (i mod 2^32, i div 2^32, 0x466F7267, 0) under key
+ * (seed mod 2^32, seed div 2^32) (Salmon et al., SC'11).  O(k) time and memory.
+ * Requires 1 <= k <= n.  Synchronous, no GPU use. */
+int skm_forgy_indices(uint64_t seed, int64_t n, int k, int64_t *idx_host);
 
 /* Haar-random orthogonal d x d matrix (HOST helper, host output P_host[d][d],
  * float32 row-major): Householder QR of a Gaussian matrix drawn with
@@ -399,8 +432,10 @@ int skm_update_finalize(const skm_data *x, const void *partial, const int64_t *c
  * STEP 2 once more for the final assignment.
  *  cfg->iters >= 0.  Initial centroids: C_init (device, per-repr layout of
  *  skm_assign) when non-NULL, else the points init_idx[0..k) (device int64,
- *  Forgy, STEP 1): F32/BF16 rows, SQ8 codes, RBQ1 / LVQ4 decoded points (the
- *  decode-average of one member).
+ *  Forgy, STEP 1): F32 rows, SQ8 codes, RBQ1 / LVQ4 decoded points (the
+ *  decode-average of one member); when init_idx is NULL too, the points
+ *  skm_forgy_indices(cfg->seed, n, k) (drawn on the host, copied to the
+ *  workspace).  BF16 points need C_init (fp32 centroids).
  *  An init_idx entry outside [0, n) makes the call fail with
  *  SKM_ERR_DEVICE_CHECK before any iteration; a tensor-core pipeline wait
  *  that exceeds its 2 s limit makes it return SKM_ERR_TIMEOUT.
@@ -414,7 +449,9 @@ typedef struct skm_fit_config {
     int32_t k;
     int32_t iters;
     int32_t empty_policy;  /* SKM_EMPTY_KEEP (0) or SKM_EMPTY_SPLIT (1), below */
-    int32_t reserved[5];
+    int32_t reserved0;
+    uint64_t seed;         /* Forgy seed, used when C_init and init_idx are NULL */
+    int32_t reserved[2];
 } skm_fit_config;
 
 /* Empty clusters after an update (Section 2.3 STEP 3: splitting large clusters
@@ -426,6 +463,59 @@ int skm_fit(const skm_fit_config *cfg, const skm_data *x, const void *C_init,
             const int64_t *init_idx, void *C_out, int32_t *assign_out, float *dist_out,
             double *objective_host, skm_stats *stats_host, void *ws, size_t ws_bytes,
             void *stream);
+
+/* ------------------------------------------------------------------------
+ * One Lloyd iteration (Section 2.3: STEP 2 then STEP 3) of points held in
+ * HOST memory, for callers whose points do not stay on the GPU: the points
+ * cross the host link once per iteration, so the call overlaps that copy with
+ * the work.  The rows are cut into cfg->chunks ranges of ceil(n / chunks)
+ * rows; range i is copied to the device on cfg->copy_stream into one of three
+ * range buffers of the workspace while `stream` assigns earlier ranges
+ * (skm_assign on a device view of the range) and adds their cluster sums into
+ * partial sums (skm_update's sharded form); a buffer is refilled once its
+ * range's assignments have been sent back.  Then cfg->exchange (if set) runs,
+ * the partial sums are finalised (skm_update_finalize) and the centroids are
+ * copied back.
+ *  x: a HOST view of the points: repr F32, BF16 or SQ8, flags 0, screen NULL,
+ *     x->x in page-locked host memory (cudaHostAlloc, cudaHostRegister or a
+ *     pinned PyTorch tensor), else SKM_ERR_INVALID_ARG before any work.
+ *  C_host (host): the centroids this iteration assigns to (per-repr layout
+ *     of skm_assign); C_host_out (host, may equal C_host): the updated
+ *     centroids; assign_host (host int32[n]): the assignments of STEP 2;
+ *     counts_host (host int64[k] or NULL): member counts; objective_host
+ *     (host double or NULL): fp64 sum of the STEP 2 distances.
+ *  cfg->copy_stream: cudaStream_t of the host-to-device copies (NULL: they go
+ *     on `stream`, without overlap).
+ *  cfg->partial / cfg->counts: device buffers for the partial sums (double
+ *     [k][d], int64 [k][d] for SQ8) and member counts (int64 [k]); NULL: taken
+ *     from the workspace.
+ *  cfg->exchange: NULL, or a host function called once all ranges are
+ *     summed with (partial, counts, cfg->user, stream) and enqueued work on
+ *     `stream` before it returns (a multi-process caller all-reduces the
+ *     partial sums and counts there: the path's one exchange per iteration);
+ *     a non-zero return ends the call with SKM_ERR_EXCHANGE.
+ *  ws: device workspace of skm_step_host_workspace_size(cfg, x) bytes (0 when
+ *     the arguments are invalid), 256-byte aligned.
+ * Synchronous: returns once the outputs are in host memory (both streams
+ * synchronised).  Results equal skm_assign followed by skm_update with
+ * partial sums and skm_update_finalize on the same points.
+ * ------------------------------------------------------------------------ */
+typedef int (*skm_exchange_fn)(void *partial, int64_t *counts, void *user, void *stream);
+typedef struct skm_step_host_config {
+    int32_t k;
+    int32_t chunks;         /* row ranges, 1..256                              */
+    void *copy_stream;
+    void *partial;
+    int64_t *counts;
+    skm_exchange_fn exchange;
+    void *user;
+    int32_t reserved[4];
+} skm_step_host_config;
+
+size_t skm_step_host_workspace_size(const skm_step_host_config *cfg, const skm_data *x);
+int skm_lloyd_step_host(const skm_step_host_config *cfg, const skm_data *x, const void *C_host,
+                        void *C_host_out, int32_t *assign_host, int64_t *counts_host,
+                        double *objective_host, void *ws, size_t ws_bytes, void *stream);
 
 /* ------------------------------------------------------------------------
  * Hierarchical k-means (Section 4, "Other Accelerators": Hierarchical k-Means): MESO-CLUSTERING

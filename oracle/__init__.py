@@ -93,6 +93,8 @@ def lib():
                 "or_lvq4_assign": ([vp, vp, i64, i32, vp, vp, vp, i32, vp, vp], None),
                 "or_lvq4_exponent": ([vp, i64], i32),
                 "or_lvq4_update": ([vp, vp, i64, i32, i32, vp, i32, vp, vp], None),
+                "or_philox4x32_10": ([vp, vp, vp], None),
+                "or_forgy_indices": ([ctypes.c_uint64, i64, i32, vp], None),
             }
             for name, (args, res) in sig.items():
                 fn = getattr(L, name)
@@ -684,3 +686,23 @@ def hierarchical(kind, data, k, m, meso_init, meso_iters, fine_iters, refine=Fal
         else:
             C, a = lloyd_rbq1(r["codes"], r["nx2"], r["F"], r["popx"], r["d"], r["m"], C, 1, r["e"])
     return C, a, am, kf
+
+
+# --------------------------------------------------------------------------
+# STEP 1 (Section 2.3): seeded Forgy initialisation
+# --------------------------------------------------------------------------
+def philox4x32_10(ctr, key):
+    """Philox4x32-10 of a 4-word counter under a 2-word key (4 uint32 words)."""
+    c = np.asarray(ctr, dtype=np.uint32)
+    k = np.asarray(key, dtype=np.uint32)
+    out = np.empty(4, np.uint32)
+    lib().or_philox4x32_10(_p(c), _p(k), _p(out))
+    return out
+
+
+def forgy_indices(seed, n, k):
+    """The first k entries of the seeded Fisher-Yates permutation of range(n)
+    (int64[k]); the draw is defined in skm_oracle.c."""
+    out = np.empty(int(k), np.int64)
+    lib().or_forgy_indices(ctypes.c_uint64(int(seed) & (2**64 - 1)), int(n), int(k), _p(out))
+    return out

@@ -875,3 +875,66 @@ void or_lvq4_update(const uint8_t *xc, const float *xfac, int64_t n, int d, int 
     free(T);
     free(U);
 }
+
+/* ------------------------------------------------------------------------ */
+/* STEP 1 (Section 2.3): Forgy initialisation from a seed -- the first k     */
+/* entries of a uniformly random permutation of 0..n-1.                      */
+/*                                                                           */
+/* Random bits: Philox4x32-10 (Salmon, Moraes, Dror, Shaw, "Parallel random  */
+/* numbers: as easy as 1, 2, 3", SC'11): ten rounds on a 4 x 32-bit counter   */
+/* under a 2 x 32-bit key; each round multiplies counter words 0 and 2 by     */
+/* 0xD2511F53 and 0xCD9E8D57 (64-bit products split into high and low        */
+/* halves) and forms (hi1 ^ c1 ^ k0, lo1, hi0 ^ c3 ^ k1, lo0); the key is     */
+/* advanced by the Weyl constants (0x9E3779B9, 0xBB67AE85) between rounds.   */
+/* Parity: pinned by the published known-answer vectors of Philox4x32-10.    */
+/* ------------------------------------------------------------------------ */
+void or_philox4x32_10(const uint32_t ctr_in[4], const uint32_t key_in[2], uint32_t out[4]) {
+    uint32_t c[4] = {ctr_in[0], ctr_in[1], ctr_in[2], ctr_in[3]};
+    uint32_t k0 = key_in[0], k1 = key_in[1];
+    for (int round = 0; round < 10; ++round) {
+        if (round > 0) {
+            k0 += 0x9E3779B9u;
+            k1 += 0xBB67AE85u;
+        }
+        uint64_t p0 = (uint64_t)0xD2511F53u * (uint64_t)c[0];
+        uint64_t p1 = (uint64_t)0xCD9E8D57u * (uint64_t)c[2];
+        uint32_t hi0 = (uint32_t)(p0 >> 32), lo0 = (uint32_t)p0;
+        uint32_t hi1 = (uint32_t)(p1 >> 32), lo1 = (uint32_t)p1;
+        uint32_t n0 = hi1 ^ c[1] ^ k0;
+        uint32_t n2 = hi0 ^ c[3] ^ k1;
+        c[0] = n0;
+        c[1] = lo1;
+        c[2] = n2;
+        c[3] = lo0;
+    }
+    out[0] = c[0];
+    out[1] = c[1];
+    out[2] = c[2];
+    out[3] = c[3];
+}
+
+/* Fisher-Yates on the identity sequence a = (0, 1, ..., n-1), positions      */
+/* i = 0 .. k-1 only: draw i is Philox4x32-10 of counter (i mod 2^32,        */
+/* i div 2^32, 0x466F7267, 0) under key (seed mod 2^32, seed div 2^32);      */
+/* r = w0 2^32 + w1; j = i + floor(r (n - i) / 2^64); swap a[i] and a[j].     */
+/* out[0..k) = a[0..k).  Parity: pinned by the permutation properties (every */
+/* index once, k = n a full permutation, uniform first entry).               */
+void or_forgy_indices(uint64_t seed, int64_t n, int k, int64_t *out) {
+    int64_t *a = (int64_t *)malloc(sizeof(int64_t) * (size_t)n);
+    for (int64_t i = 0; i < n; ++i) a[i] = i;
+    const uint32_t key[2] = {(uint32_t)seed, (uint32_t)(seed >> 32)};
+    for (int64_t i = 0; i < k; ++i) {
+        const uint32_t ctr[4] = {(uint32_t)i, (uint32_t)((uint64_t)i >> 32), 0x466F7267u, 0u};
+        uint32_t w[4];
+        or_philox4x32_10(ctr, key, w);
+        const uint64_t r = ((uint64_t)w[0] << 32) | (uint64_t)w[1];
+        const uint64_t span = (uint64_t)(n - i);
+        const uint64_t off = (uint64_t)(((unsigned __int128)r * span) >> 64);
+        const int64_t j = i + (int64_t)off;
+        const int64_t t = a[i];
+        a[i] = a[j];
+        a[j] = t;
+        out[i] = a[i];
+    }
+    free(a);
+}

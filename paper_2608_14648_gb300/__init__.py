@@ -41,7 +41,8 @@ EXPORTED_SYMBOLS = [
     "skm_assign_segmented",
     "skm_update",
     "skm_merge_partials", "skm_update_finalize", "skm_fit", "skm_split_empty", "skm_hier_workspace_size",
-    "skm_fit_hierarchical", "skm_objective", "skm_sq8_decode",
+    "skm_fit_hierarchical", "skm_objective", "skm_sq8_decode", "skm_step_host_workspace_size",
+    "skm_lloyd_step_host", "skm_inject_fault", "skm_fault_armed", "skm_forgy_indices",
 ]
 
 
@@ -83,7 +84,18 @@ class HierConfig(ctypes.Structure):
 
 class FitConfig(ctypes.Structure):
     _fields_ = [("k", ctypes.c_int32), ("iters", ctypes.c_int32), ("empty_policy", ctypes.c_int32),
-                ("reserved", ctypes.c_int32 * 5)]
+                ("reserved0", ctypes.c_int32), ("seed", ctypes.c_uint64), ("reserved", ctypes.c_int32 * 2)]
+
+
+EXCHANGE_FN = ctypes.CFUNCTYPE(ctypes.c_int, ctypes.c_void_p, ctypes.c_void_p, ctypes.c_void_p, ctypes.c_void_p)
+
+
+class StepHostConfig(ctypes.Structure):
+    """skm_step_host_config (include/skm.h)."""
+
+    _fields_ = [("k", ctypes.c_int32), ("chunks", ctypes.c_int32), ("copy_stream", ctypes.c_void_p),
+                ("partial", ctypes.c_void_p), ("counts", ctypes.c_void_p), ("exchange", EXCHANGE_FN),
+                ("user", ctypes.c_void_p), ("reserved", ctypes.c_int32 * 4)]
 
 
 def lib_path() -> str:
@@ -107,6 +119,7 @@ def lib():
             "skm_screen_prep": ([vp, vp, sz, vp], i32),
             "skm_project": ([vp, i64, i32, vp, vp, i32, i32, vp, vp, sz, vp], i32),
             "skm_make_rotation": ([u64, i32, vp], i32),
+            "skm_forgy_indices": ([u64, i64, i32, vp], i32),
             "skm_project_hadamard": ([vp, i64, i32, vp, vp, i32, i32, vp, vp], i32),
             "skm_unproject": ([vp, i64, i32, vp, vp, i32, vp, vp], i32),
             "skm_copy_from_host": ([vp, vp, sz, vp], i32),
@@ -126,6 +139,10 @@ def lib():
             "skm_fit_hierarchical": ([vp, vp, vp, vp, vp, vp, vp, vp, vp, sz, vp], i32),
             "skm_objective": ([vp, i32, i64, i32, vp, i32, vp, vp, vp, sz, vp], i32),
             "skm_sq8_decode": ([vp, i64, i32, vp, vp, vp, vp], i32),
+            "skm_inject_fault": ([i32, i32], i32),
+            "skm_fault_armed": ([i32], i32),
+            "skm_step_host_workspace_size": ([vp, vp], sz),
+            "skm_lloyd_step_host": ([vp, vp, vp, vp, vp, vp, vp, vp, sz, vp], i32),
         }
         for name, (args, res) in sig.items():
             fn = getattr(L, name)
@@ -436,9 +453,17 @@ def skm_split_empty(pts: Points, C_inout, counts, stream=None):
     return C_inout
 
 
+def skm_forgy_indices(seed, n, k):
+    """Seeded Forgy indices (int64 CPU tensor [k]); see include/skm.h."""
+    out = torch.empty(int(k), dtype=torch.int64)
+    _check(lib().skm_forgy_indices(int(seed) & (2**64 - 1), int(n), int(k), ctypes.c_void_p(out.data_ptr())))
+    return out
+
+
 def skm_fit(pts: Points, k, iters, C_init=None, init_idx=None, want_objective=True, want_dist=True,
-            ws=None, stream=None, empty_policy=EMPTY_KEEP):
-    """Returns (C, assign, dist or None, objective list or None, stats dict)."""
+            ws=None, stream=None, empty_policy=EMPTY_KEEP, seed=0):
+    """Returns (C, assign, dist or None, objective list or None, stats dict).
+    With neither C_init nor init_idx the library draws Forgy indices from `seed`."""
     dev = pts.device
     if ws is None:
         ws = _ws(skm_workspace_size(OP_FIT, pts, k), dev)
@@ -450,7 +475,7 @@ def skm_fit(pts: Points, k, iters, C_init=None, init_idx=None, want_objective=Tr
     dist = torch.empty(pts.n, device=dev, dtype=torch.float32) if want_dist else None
     obj = (ctypes.c_double * (iters + 1))() if want_objective else None
     st = Stats()
-    cfg = FitConfig(int(k), int(iters), int(empty_policy))
+    cfg = FitConfig(int(k), int(iters), int(empty_policy), 0, int(seed) & (2**64 - 1))
     _check(lib().skm_fit(ctypes.byref(cfg), ctypes.byref(pts.ref), _ptr(C_init), _ptr(init_idx), _ptr(C),
                          _ptr(assign), _ptr(dist), obj, ctypes.byref(st), _ptr(ws), ws.numel(), _stream(stream)))
     stats = {"rescored_rows": st.rescored_rows, "fallback_rows": st.fallback_rows,
@@ -499,3 +524,73 @@ def skm_sq8_decode(codes, b, s, stream=None):
     Y = torch.empty(n, d, device=codes.device, dtype=torch.float32)
     _check(lib().skm_sq8_decode(_ptr(codes), n, d, _ptr(b), _ptr(s), _ptr(Y), _stream(stream)))
     return Y
+
+
+def _host_data(repr_, X_host, d):
+    if X_host.device.type != "cpu" or not X_host.is_contiguous():
+        raise ValueError("points: a contiguous host tensor")
+    return Data(repr_, int(d), X_host.shape[0], X_host.data_ptr(), None, None, None, None, 0, 0, None, None)
+
+
+class LloydStepHost:
+    """skm_lloyd_step_host with its workspace: one Lloyd iteration of points
+    held in (pinned) host memory per call.  `exchange` (optional) is a
+    callable run between the partial sums and the finalisation; it must
+    enqueue its work on the step's stream and then reads/writes the tensors
+    `self.partial` and `self.counts`."""
+
+    def __init__(self, repr_, X_host, d, k, chunks=16, device=None, copy_stream=None, exchange=None):
+        self.device = torch.device("cuda") if device is None else torch.device(device)
+        self.repr, self.k, self.d = repr_, int(k), int(d)
+        self.X_host = X_host
+        self.ref = _host_data(repr_, X_host, d)
+        pdt = torch.int64 if repr_ == REPR_SQ8 else torch.float64
+        self.partial = torch.zeros(self.k, self.d, dtype=pdt, device=self.device)
+        self.counts = torch.zeros(self.k, dtype=torch.int64, device=self.device)
+        self.copy_stream = copy_stream if copy_stream is not None else torch.cuda.Stream(self.device)
+        self._user_exchange = exchange
+        self._cb = EXCHANGE_FN(self._exchange) if exchange is not None else EXCHANGE_FN()
+        self.cfg = StepHostConfig(self.k, int(chunks), ctypes.c_void_p(self.copy_stream.cuda_stream),
+                                  self.partial.data_ptr(), self.counts.data_ptr(), self._cb, None)
+        nbytes = lib().skm_step_host_workspace_size(ctypes.byref(self.cfg), ctypes.byref(self.ref))
+        if nbytes == 0:
+            raise SkmError(1, lib().skm_last_error().decode())
+        self.ws = _ws(nbytes, self.device)
+
+    def _exchange(self, partial, counts, user, stream):
+        # the hook's work goes on the stream this step was called with (the
+        # library passes that stream's handle; a handle of 0 is the default
+        # stream, which torch.cuda.ExternalStream(0) would not give back)
+        try:
+            with torch.cuda.stream(self._call_stream):
+                self._user_exchange()
+            return 0
+        except Exception:  # reported to the library as a failed exchange
+            return 1
+
+    def __call__(self, C_host, C_host_out=None, assign_host=None, counts_host=None, want_objective=False,
+                 stream=None):
+        """Returns (C_host_out, assign_host, counts_host or None, objective or None)."""
+        n = self.X_host.shape[0]
+        C_host_out = C_host if C_host_out is None else C_host_out
+        if assign_host is None:
+            assign_host = torch.empty(n, dtype=torch.int32, pin_memory=True)
+        obj = ctypes.c_double(0.0) if want_objective else None
+        self._call_stream = stream if stream is not None else torch.cuda.current_stream(self.device)
+        _check(lib().skm_lloyd_step_host(ctypes.byref(self.cfg), ctypes.byref(self.ref), _ptr(C_host),
+                                         _ptr(C_host_out), _ptr(assign_host), _ptr(counts_host),
+                                         ctypes.byref(obj) if obj is not None else None, _ptr(self.ws),
+                                         self.ws.numel(), _stream(self._call_stream)))
+        return C_host_out, assign_host, counts_host, (obj.value if obj is not None else None)
+
+
+FAULT_WORKSPACE, FAULT_LAUNCH, FAULT_STATUS, FAULT_WAIT = 1, 2, 3, 4
+
+
+def skm_inject_fault(kind, count=1):
+    """Arms `count` occurrences of an SKM_FAULT_* (0 disarms); see include/skm.h."""
+    _check(lib().skm_inject_fault(int(kind), int(count)))
+
+
+def skm_fault_armed(kind) -> int:
+    return int(lib().skm_fault_armed(int(kind)))

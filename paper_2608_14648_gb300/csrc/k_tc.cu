@@ -149,6 +149,10 @@ struct TcParams {
     void *y;
     int y_bf16;
     int ydout;
+    // Fault injection (0 = off): the producer first waits this long on a
+    // barrier that nothing arrives on, so the launch gives up before it has
+    // loaded anything and reports through the abort flag.
+    unsigned long long inject_wait_ns;
 };
 
 // ------------------------------------------------------------- PTX helpers
@@ -183,18 +187,29 @@ __device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
 }
 // Bounded wait: false when the abort flag is raised or the limit elapses
 // (the flag is then raised so that every role stops).
-__device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, volatile int32_t *abort_flag) {
+__device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, volatile int32_t *abort_flag,
+                                          unsigned long long limit_ns = WAIT_LIMIT_NS) {
     if (mbar_try_wait(bar, parity)) return true;
     const unsigned long long t0 = globaltimer();
     for (uint32_t i = 1;; ++i) {
         if (mbar_try_wait(bar, parity)) return true;
         if ((i & 255) == 0) {
             if (*abort_flag) return false;
-            if (globaltimer() - t0 > WAIT_LIMIT_NS) {
+            if (globaltimer() - t0 > limit_ns) {
                 *abort_flag = 1;
                 return false;
             }
         }
+    }
+}
+// Wait with the limit only (the abort flag is already up): used after a
+// role gave up, to let the asynchronous copies or MMAs it had issued finish
+// before the CTA releases its shared memory and TMEM.
+__device__ __forceinline__ bool mbar_drain(uint32_t bar, uint32_t parity) {
+    const unsigned long long t0 = globaltimer();
+    for (uint32_t i = 0;; ++i) {
+        if (mbar_try_wait(bar, parity)) return true;
+        if ((i & 255) == 255 && globaltimer() - t0 > WAIT_LIMIT_NS) return false;
     }
 }
 __device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap *map, int x, int y,
@@ -428,6 +443,10 @@ __global__ void __launch_bounds__(tc_threads<NH>(), 1)
     auto tfull_bar = [&](int b) { return bar0 + 8u * (2 * STAGES + b); };
     auto tempty_bar = [&](int b) { return bar0 + 8u * (2 * STAGES + 2 + b); };
     uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(bars + 2 * STAGES + 4);
+    // two more barriers after the TMEM slot: the MMA warp's drain on abort and
+    // the injected wait (nothing arrives on either otherwise)
+    const uint32_t drain_bar = bar0 + 8u * (2 * STAGES + 5);
+    const uint32_t inject_bar = bar0 + 8u * (2 * STAGES + 6);
     // the epilogue's merge buffer starts 256 bytes after tmem_slot (see tc_smem_bytes)
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -444,6 +463,8 @@ __global__ void __launch_bounds__(tc_threads<NH>(), 1)
             mbar_init(tfull_bar(b), 1);
             mbar_init(tempty_bar(b), epi_threads<NH>() / NS);
         }
+        mbar_init(drain_bar, 1);
+        mbar_init(inject_bar, 1);
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
         asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmA)) : "memory");
         asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmB)) : "memory");
@@ -512,6 +533,8 @@ __global__ void __launch_bounds__(tc_threads<NH>(), 1)
     if (warp == 0) {
         if (lane == 0) {  // ---------------------------------------- TMA producer
             uint32_t it = 0;
+            if (p.inject_wait_ns && !mbar_wait(inject_bar, 0u, abort_flag, p.inject_wait_ns)) goto producer_done;
+            {
             JobStream js[NS];
             for (int s = 0; s < NS; ++s) {
                 js[s].g = g0 + s * gstep;
@@ -538,11 +561,20 @@ __global__ void __launch_bounds__(tc_threads<NH>(), 1)
                     }
                 }
             }
-        producer_done:;
+            }
+        producer_done:
+            // Every stage fill issued so far lands before the CTA can exit (after
+            // a normal run the MMA warp has consumed them all and this returns at
+            // once; after an abort it waits for the copies still in flight).
+            for (uint32_t s = 0; s < (uint32_t)STAGES && s < it; ++s) {
+                const uint32_t last = s + ((it - 1u - s) / STAGES) * STAGES;
+                mbar_drain(full_bar(s), (last / STAGES) & 1u);
+            }
         }
     } else if (warp == 1) {
         if (lane == 0) {  // ---------------------------------------- MMA issuer
             uint32_t it = 0, job = 0;
+            bool issued = false, gave_up = true;
             uint32_t jc[NS];
             JobStream js[NS];
             for (int s = 0; s < NS; ++s) {
@@ -580,12 +612,20 @@ __global__ void __launch_bounds__(tc_threads<NH>(), 1)
                             else
                                 tc_mma(dcol, ad + 2u * kk, bd + 2u * kk, IDESC, (kc | kk) != 0);
                         }
+                        issued = true;
                         tc_commit(empty_bar(s));
                     }
                     tc_commit(tfull_bar(b));
                 }
             }
-        mma_done:;
+            gave_up = false;
+        mma_done:
+            // After an abort, the MMAs issued so far complete before TMEM is
+            // released (after a normal run the epilogue has waited for them all).
+            if (gave_up && issued) {
+                tc_commit(drain_bar);
+                mbar_drain(drain_bar, 0u);
+            }
         }
     } else {  // ------------------------------------------------------- epilogue
         constexpr int NHG = NH / NS;     // warps per TMEM lane quarter in a group
@@ -1530,6 +1570,7 @@ int launch_tc_kind(const void *xs, int64_t n, int dp, int d, const void *cs, int
     p.k = k;
     p.nct = (int)cdiv(k, BN);
     p.nkc = (int)cdiv(d, 128 / eb);
+    p.inject_wait_ns = fault_take(SKM_FAULT_WAIT) ? 1000000ull : 0ull;  // 1 ms
     const int grid = (int)std::min<int64_t>(device_sms(), p.nrt);
     kern<<<grid, tc_threads<NH>(), SMEM, st>>>(ma, mb, p);
     SKM_CUDA_TRY(launched());

@@ -3,10 +3,13 @@
 // Lloyd k-means hot path (Section 2.3) for each representation.
 #include <stdarg.h>
 #include <stdio.h>
+#include <stdlib.h>
+#include <string.h>
 
 #include <algorithm>
 #include <atomic>
 #include <cmath>
+#include <mutex>
 #include <vector>
 
 #include "skm_internal.cuh"
@@ -17,9 +20,32 @@ namespace skm {
 static thread_local char g_err[512] = "";
 static std::atomic<unsigned long long> g_launches{0};
 
+// ---- fault injection (host side; SKM_FAULT_* kinds 1..4)
+static std::atomic<int> g_fault[5];
+static std::once_flag g_fault_env;
+
+static void fault_from_env() {
+    const char *v = getenv("SKM_FAULT");
+    if (!v) return;
+    const char *names[5] = {"", "workspace", "launch", "status", "wait"};
+    for (int kind = 1; kind <= 4; ++kind)
+        if (strcmp(v, names[kind]) == 0) g_fault[kind].store(1);
+}
+
+bool fault_take(int kind) {
+    std::call_once(g_fault_env, fault_from_env);
+    if (kind < 1 || kind > 4) return false;
+    int c = g_fault[kind].load();
+    while (c > 0)
+        if (g_fault[kind].compare_exchange_weak(c, c - 1)) return true;
+    return false;
+}
+
 cudaError_t launched(int count) {
     g_launches.fetch_add((unsigned long long)count, std::memory_order_relaxed);
-    return cudaGetLastError();
+    const cudaError_t e = cudaGetLastError();
+    if (e == cudaSuccess && fault_take(SKM_FAULT_LAUNCH)) return cudaErrorLaunchFailure;
+    return e;
 }
 
 int set_error(int code, const char *fmt, ...) {
@@ -174,6 +200,7 @@ struct FitBufs {
     int *e_dev = nullptr;
     int *status = nullptr;
     int64_t *counts = nullptr;
+    int64_t *init_idx = nullptr;
 };
 
 static void plan_fit(const skm_data *x, int k, Carver &cv, FitBufs &b) {
@@ -194,9 +221,12 @@ static void plan_fit(const skm_data *x, int k, Carver &cv, FitBufs &b) {
     b.e_dev = cv.take<int>(1);
     b.status = cv.take<int>(1);
     b.counts = cv.take<int64_t>(k);
+    b.init_idx = cv.take<int64_t>(k);  // seeded Forgy indices (host-drawn)
 }
 
 static int need_ws(const Carver &cv, size_t ws_bytes, void *ws) {
+    if (fault_take(SKM_FAULT_WORKSPACE))
+        return set_error(SKM_ERR_NO_MEMORY, "injected fault: workspace reported too small");
     if (cv.off > ws_bytes)
         return set_error(SKM_ERR_NO_MEMORY, "workspace too small: need %zu bytes, got %zu", cv.off,
                          ws_bytes);
@@ -344,6 +374,18 @@ extern "C" {
 
 const char *skm_last_error(void) { return g_err; }
 
+int skm_inject_fault(int kind, int count) {
+    std::call_once(g_fault_env, fault_from_env);
+    if (kind < 1 || kind > 4 || count < 0) return set_error(SKM_ERR_INVALID_ARG, "fault kind %d, count %d", kind, count);
+    g_fault[kind].store(count);
+    return SKM_OK;
+}
+
+int skm_fault_armed(int kind) {
+    std::call_once(g_fault_env, fault_from_env);
+    return (kind < 1 || kind > 4) ? 0 : g_fault[kind].load();
+}
+
 int skm_version(void) { return 100; }
 
 uint64_t skm_kernel_launches(void) { return (uint64_t)g_launches.load(std::memory_order_relaxed); }
@@ -465,6 +507,13 @@ int skm_copy_from_host(void *dst, const void *src_host, size_t bytes, void *stre
                          cudaGetErrorString(e));
     }
     SKM_CUDA_TRY(launch_copy_from_host(src_dev, dst, bytes, S(stream)));
+    return SKM_OK;
+}
+
+int skm_forgy_indices(uint64_t seed, int64_t n, int k, int64_t *idx_host) {
+    if (!idx_host) return set_error(SKM_ERR_INVALID_ARG, "idx_host is NULL");
+    if (n < 1 || k < 1 || (int64_t)k > n) return set_error(SKM_ERR_INVALID_ARG, "need 1 <= k <= n (k=%d n=%lld)", k, (long long)n);
+    forgy_indices(seed, n, k, idx_host);
     return SKM_OK;
 }
 
@@ -974,8 +1023,8 @@ int skm_fit(const skm_fit_config *cfg, const skm_data *x, const void *C_init,
     if (cfg->empty_policy != SKM_EMPTY_KEEP && cfg->empty_policy != SKM_EMPTY_SPLIT)
         return set_error(SKM_ERR_INVALID_ARG, "empty_policy = %d", cfg->empty_policy);
     if (!C_out || !assign_out) return set_error(SKM_ERR_INVALID_ARG, "C_out and assign_out required");
-    if (!C_init && !init_idx)
-        return set_error(SKM_ERR_INVALID_ARG, "one of C_init / init_idx is required");
+    if (!C_init && x->repr == SKM_REPR_BF16)
+        return set_error(SKM_ERR_INVALID_ARG, "BF16 fit needs fp32 C_init");
     cudaStream_t st = S(stream);
     Carver cv(ws, ws_bytes);
     FitBufs b;
@@ -1004,7 +1053,16 @@ int skm_fit(const skm_fit_config *cfg, const skm_data *x, const void *C_init,
         SKM_CUDA_TRY(cudaStreamSynchronize(st));
         xd.rbq1_exp = e;
     }
-    // STEP 1: initial centroids
+    // STEP 1: initial centroids (Forgy from cfg->seed when neither C_init
+    // nor init_idx is given)
+    std::vector<int64_t> seeded;
+    if (!C_init && !init_idx) {
+        seeded.resize(k);
+        forgy_indices(cfg->seed, n, k, seeded.data());
+        SKM_CUDA_TRY(cudaMemcpyAsync(b.init_idx, seeded.data(), sizeof(int64_t) * (size_t)k, cudaMemcpyHostToDevice,
+                                     st));
+        init_idx = b.init_idx;
+    }
     SKM_CUDA_TRY(cudaMemsetAsync(b.status, 0, sizeof(int), st));
     SKM_CUDA_TRY(cudaMemsetAsync(b.u.flag, 0, sizeof(int32_t), st));
     if (C_init) {
@@ -1049,7 +1107,13 @@ int skm_fit(const skm_fit_config *cfg, const skm_data *x, const void *C_init,
             SKM_CUDA_TRY(launch_split_empty(C_out, x->repr == SKM_REPR_SQ8 ? 1 : 4, b.counts, k, x->d,
                                             b.u.wsplit, st));
     }
-    SKM_CUDA_TRY(cudaStreamSynchronize(st));
+    if (fault_take(SKM_FAULT_STATUS)) SKM_CUDA_TRY(cudaMemsetAsync(b.status, 0xff, sizeof(int), st));
+    {
+        int bad = 0;
+        SKM_CUDA_TRY(cudaMemcpyAsync(&bad, b.status, sizeof(int), cudaMemcpyDeviceToHost, st));
+        SKM_CUDA_TRY(cudaStreamSynchronize(st));
+        if (bad) return set_error(SKM_ERR_DEVICE_CHECK, "the device status word is set (%d)", bad);
+    }
     skm_stats local;
     memset(&local, 0, sizeof(local));
     SKM_TRY(tc_read_stats(b.a.tc, &local, st));

@@ -33,6 +33,9 @@ int set_error(int code, const char *fmt, ...);
 // Counts `count` kernel launches (host-side, process-wide) and returns
 // cudaGetLastError(); every launcher returns through it.
 cudaError_t launched(int count = 1);
+// True (and one armed occurrence used up) when an SKM_FAULT_* of this kind
+// is armed (skm_inject_fault or the SKM_FAULT environment variable).
+bool fault_take(int kind);
 
 // ---- workspace carving ------------------------------------------------------
 // Sub-buffers are carved from the caller's workspace at 256-byte boundaries.
@@ -306,6 +309,7 @@ cudaError_t launch_lvq4_decode_rows(const uint32_t *codes, const float4 *fac, in
 
 // host helpers (skm_linalg.cpp)
 void philox_gaussians(uint64_t seed, int64_t count, double *out);
+void forgy_indices(uint64_t seed, int64_t n, int k, int64_t *out);
 void householder_qr_q(int d, double *A /* d*d in, Q out, row-major */);
 int symmetric_eigen(int n, double *A /* in: symmetric; out: eigenvectors as columns */,
                     double *w /* eigenvalues */);

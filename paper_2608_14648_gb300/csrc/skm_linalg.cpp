@@ -12,6 +12,7 @@
 #include <string.h>
 
 #include <algorithm>
+#include <unordered_map>
 #include <vector>
 
 namespace skm {
@@ -50,6 +51,31 @@ void philox_gaussians(uint64_t seed, int64_t count, double *out) {
         const double rad = sqrt(-2.0 * log(u1));
         out[2 * blk] = rad * cos(two_pi * u2);
         if (2 * blk + 1 < count) out[2 * blk + 1] = rad * sin(two_pi * u2);
+    }
+}
+
+// Forgy (Section 2.3 STEP 1) from a seed: positions 0..k-1 of a Fisher-Yates
+// shuffle of (0, 1, ..., n-1); draw i = Philox4x32-10 of counter (i lo, i hi,
+// 0x466F7267, 0) under key (seed lo, seed hi), r = w0 2^32 + w1, and position
+// i swaps with i + floor(r (n - i) / 2^64).  Only the displaced positions are
+// stored (a hash map), so the work and memory are O(k) whatever n is.
+void forgy_indices(uint64_t seed, int64_t n, int k, int64_t *out) {
+    const uint32_t k0 = (uint32_t)seed, k1 = (uint32_t)(seed >> 32);
+    std::unordered_map<int64_t, int64_t> moved;
+    moved.reserve((size_t)k * 2 + 16);
+    auto at = [&](int64_t p) {
+        auto it = moved.find(p);
+        return it == moved.end() ? p : it->second;
+    };
+    for (int64_t i = 0; i < k; ++i) {
+        uint32_t c[4] = {(uint32_t)i, (uint32_t)((uint64_t)i >> 32), 0x466F7267u, 0u};
+        philox4x32_10(c, k0, k1);
+        const uint64_t r = ((uint64_t)c[0] << 32) | c[1];
+        const int64_t j = i + (int64_t)(((unsigned __int128)r * (uint64_t)(n - i)) >> 64);
+        const int64_t vi = at(i), vj = at(j);
+        moved[j] = vi;
+        moved[i] = vj;
+        out[i] = vj;
     }
 }
 

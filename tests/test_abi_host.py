@@ -72,10 +72,11 @@ def test_invalid_arguments_are_rejected_before_launch(skm):
     rc = L.skm_assign(ctypes.byref(_data(skm, repr_=1)), FAKE, 4, None, FAKE, None, ctypes.c_void_p(0x1010), need,
                       None)
     assert rc == 1
-    # fit without any initialisation
+    # BF16 fit without fp32 initial centroids (seeded Forgy cannot build them)
     cfg = skm.FitConfig(4, 3)
-    rc = L.skm_fit(ctypes.byref(cfg), ctypes.byref(x), None, None, FAKE, FAKE, None, None, None, FAKE, 1 << 30, None)
-    assert rc == 1
+    xb = _data(skm, repr_=3)
+    rc = L.skm_fit(ctypes.byref(cfg), ctypes.byref(xb), None, None, FAKE, FAKE, None, None, None, FAKE, 1 << 30, None)
+    assert rc == 1 and b"C_init" in L.skm_last_error()
     # projection to more dims than the input
     assert L.skm_project(FAKE, 10, 8, None, FAKE, 9, 0, FAKE, None, 0, None) == 1
     # misaligned projection workspace
@@ -161,3 +162,92 @@ def test_copy_from_host_arguments(skm):
     assert L.skm_copy_from_host(None, FAKE, 16, None) == 1
     assert L.skm_copy_from_host(FAKE, None, 16, None) == 1
     assert "NULL" in L.skm_last_error().decode()
+
+
+def test_step_host_arguments_are_rejected_before_any_work(skm):
+    """skm_lloyd_step_host / skm_step_host_workspace_size: bad configurations
+    return their status (and size 0) before any CUDA call."""
+    L = skm.lib()
+    X = np.zeros((100, 16), np.float32)
+    x = skm.Data(0, 16, 100, X.ctypes.data, None, None, None, None, 0, 0)
+
+    def cfg(k=10, chunks=4):
+        return skm.StepHostConfig(k, chunks, None, None, None, skm.EXCHANGE_FN(), None)
+
+    assert L.skm_step_host_workspace_size(ctypes.byref(cfg()), ctypes.byref(x)) > 0
+    for c, code, what in [(cfg(k=101), 1, b"k = 101"), (cfg(k=0), 1, b"k = 0"), (cfg(chunks=0), 1, b"chunks"),
+                          (cfg(chunks=257), 1, b"chunks")]:
+        assert L.skm_step_host_workspace_size(ctypes.byref(c), ctypes.byref(x)) == 0
+        rc = L.skm_lloyd_step_host(ctypes.byref(c), ctypes.byref(x), FAKE, FAKE, FAKE, None, None, FAKE, 1 << 30,
+                                   None)
+        assert rc == code and what in L.skm_last_error()
+    for repr_ in (2, 4):  # RBQ1 / LVQ4: factors would need copying too
+        xr = skm.Data(repr_, 16, 100, X.ctypes.data, None, None, None, None, 0, 0)
+        assert L.skm_lloyd_step_host(ctypes.byref(cfg()), ctypes.byref(xr), FAKE, FAKE, FAKE, None, None, FAKE,
+                                     1 << 30, None) == 2
+    xf = skm.Data(0, 16, 100, X.ctypes.data, None, None, None, None, 0, 1)  # a flag
+    assert L.skm_lloyd_step_host(ctypes.byref(cfg()), ctypes.byref(xf), FAKE, FAKE, FAKE, None, None, FAKE,
+                                 1 << 30, None) == 2
+    # missing outputs / workspace
+    assert L.skm_lloyd_step_host(ctypes.byref(cfg()), ctypes.byref(x), FAKE, FAKE, None, None, None, FAKE,
+                                 1 << 30, None) == 1
+    assert L.skm_lloyd_step_host(ctypes.byref(cfg()), ctypes.byref(x), FAKE, FAKE, FAKE, None, None, None,
+                                 1 << 30, None) == 1
+    # too small a workspace
+    assert L.skm_lloyd_step_host(ctypes.byref(cfg()), ctypes.byref(x), FAKE, FAKE, FAKE, None, None,
+                                 ctypes.c_void_p(0x100000), 1024, None) == 4
+
+
+def test_fault_injection_switch(skm):
+    """skm_inject_fault arms occurrences that the first checks use up: an
+    armed workspace fault makes a valid call return SKM_ERR_NO_MEMORY before
+    anything is enqueued (so the fake pointers are never touched)."""
+    L = skm.lib()
+    assert L.skm_inject_fault(9, 1) == 1 and L.skm_inject_fault(1, -1) == 1
+    assert L.skm_fault_armed(9) == 0
+    x = _data(skm)
+    try:
+        assert L.skm_inject_fault(1, 2) == 0 and L.skm_fault_armed(1) == 2
+        for left in (1, 0):
+            rc = L.skm_assign(ctypes.byref(x), FAKE, 4, None, FAKE, None, FAKE, 1 << 30, None)
+            assert rc == 4 and b"injected" in L.skm_last_error()
+            assert L.skm_fault_armed(1) == left
+        assert L.skm_inject_fault(2, 5) == 0 and L.skm_inject_fault(2, 0) == 0 and L.skm_fault_armed(2) == 0
+    finally:
+        for kind in (1, 2, 3, 4):
+            L.skm_inject_fault(kind, 0)
+
+
+def test_fault_injection_from_environment(skm):
+    """SKM_FAULT=workspace arms one occurrence when the library first checks."""
+    import subprocess
+    import sys
+
+    code = (
+        "import ctypes, paper_2608_14648_gb300 as skm\n"
+        "L = skm.lib()\n"
+        "x = skm.Data(0, 16, 100, 0x1000, None, None, None, None, 0, 0)\n"
+        "F = ctypes.c_void_p(0x1000)\n"
+        "assert L.skm_fault_armed(1) == 1\n"
+        "assert L.skm_assign(ctypes.byref(x), F, 4, None, F, None, F, 1 << 30, None) == 4\n"
+        "assert L.skm_fault_armed(1) == 0\n"
+        "print('ok')\n")
+    env = dict(os.environ, SKM_FAULT="workspace")
+    r = subprocess.run([sys.executable, "-c", code], cwd=ROOT, env=env, capture_output=True, text=True, timeout=120)
+    assert r.returncode == 0 and r.stdout.strip() == "ok", r.stderr
+
+
+def test_forgy_indices_match_the_oracle(skm):
+    """The library's seeded Forgy draw (hash-map Fisher-Yates) equals the
+    oracle's (full-array Fisher-Yates) for the same seed: bit-exact."""
+    import oracle
+
+    L = skm.lib()
+    for seed, n, k in [(0, 10, 10), (1, 1, 1), (7, 1000, 999), (2**40 + 3, 20_000, 100),
+                       (0, 10_000_000, 10_000), (2**64 - 1, 1_000_000, 1000)]:
+        got = skm.skm_forgy_indices(seed, n, k).numpy()
+        np.testing.assert_array_equal(got, oracle.forgy_indices(seed, n, k))
+    out = np.empty(4, np.int64)
+    assert L.skm_forgy_indices(0, 3, 4, out.ctypes.data) == 1  # k > n
+    assert L.skm_forgy_indices(0, 3, 0, out.ctypes.data) == 1
+    assert L.skm_forgy_indices(0, 3, 2, None) == 1

@@ -1037,3 +1037,18 @@ def test_fit_rbq1_symmetric_trajectory_bitexact(skm):
     Co, ao = oracle.lloyd_rbq1_sym(h["codes"], h["nx2"], h["F"], h["popx"], d, h["m"], C0, iters, pts.rbq1_exp)
     np.testing.assert_array_equal(a.cpu().numpy(), ao)
     np.testing.assert_array_equal(C.cpu().numpy(), Co)
+
+
+def test_fit_seeded_forgy_matches_oracle(skm):
+    """skm_fit with neither C_init nor init_idx draws its Forgy points from
+    the seed (STEP 1); the oracle draws its own from the same seed, and the
+    SQ8 trajectories from them are bit-exact."""
+    n, d, k, iters, seed = 9001, 48, 37, 4, 2**33 + 5
+    X = _points(n, d, seed=71)
+    q = skm.skm_quantize(skm.REPR_SQ8, X.to(DEV))
+    codes = q["codes"].cpu().numpy()
+    C, a, _, _, _ = skm.skm_fit(skm.Points(skm.REPR_SQ8, q["codes"], d), k, iters, seed=seed)
+    idx = oracle.forgy_indices(seed, n, k)
+    Co, ao = oracle.lloyd_sq8(codes, codes[idx], iters)
+    np.testing.assert_array_equal(a.cpu().numpy(), ao)
+    np.testing.assert_array_equal(C.cpu().numpy(), Co)

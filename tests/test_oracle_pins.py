@@ -892,3 +892,45 @@ def test_objective_bf16_is_wcss_of_decoded_rows():
     D = cdist(oracle.bf16_to_f32(Xb).astype(np.float64), C.astype(np.float64), "sqeuclidean")
     want = float(D[np.arange(n), a].sum())
     assert math.isclose(oracle.objective_bf16(Xb, C, a), want, rel_tol=1e-12)
+
+
+# ------------------------------------------------------- seeded Forgy (STEP 1)
+def test_philox4x32_10_known_answer_vectors():
+    """The published known-answer vectors of Philox4x32-10 (Salmon et al.,
+    SC'11; the Random123 distribution's kat_vectors)."""
+    kat = [((0, 0, 0, 0), (0, 0), (0x6627E8D5, 0xE169C58D, 0xBC57AC4C, 0x9B00DBD8)),
+           ((0xFFFFFFFF,) * 4, (0xFFFFFFFF,) * 2, (0x408F276D, 0x41C83B0E, 0xA20BC7C6, 0x6D5451FD)),
+           ((0x243F6A88, 0x85A308D3, 0x13198A2E, 0x03707344), (0xA4093822, 0x299F31D0),
+            (0xD16CFE09, 0x94FDCCEB, 0x5001E420, 0x24126EA1))]
+    for ctr, key, want in kat:
+        assert tuple(int(v) for v in oracle.philox4x32_10(ctr, key)) == want
+
+
+def test_forgy_indices_are_a_permutation_prefix():
+    for seed in (0, 1, 2**40 + 7):
+        full = oracle.forgy_indices(seed, 1000, 1000)
+        assert sorted(full.tolist()) == list(range(1000))  # k = n: a permutation
+        part = oracle.forgy_indices(seed, 1000, 37)
+        np.testing.assert_array_equal(part, full[:37])  # a prefix of the same permutation
+    a = oracle.forgy_indices(5, 10_000_000, 1000)
+    assert len(set(a.tolist())) == 1000 and a.min() >= 0 and a.max() < 10_000_000
+    assert not np.array_equal(oracle.forgy_indices(6, 10_000_000, 1000), a)
+    assert oracle.forgy_indices(9, 1, 1).tolist() == [0]
+
+
+def test_forgy_indices_are_uniform():
+    """First and second entries over 20,000 seeds with n = 10: every value
+    (and every ordered pair) about equally often (chi-square)."""
+    from scipy.stats import chisquare
+
+    n, trials = 10, 20_000
+    first = np.empty(trials, np.int64)
+    second = np.empty(trials, np.int64)
+    for s in range(trials):
+        f = oracle.forgy_indices(s, n, 2)
+        first[s], second[s] = f
+    assert np.all(first != second)
+    assert chisquare(np.bincount(first, minlength=n)).pvalue > 1e-4
+    pairs = np.bincount(first * n + second, minlength=n * n).reshape(n, n)
+    off = pairs[~np.eye(n, dtype=bool)]
+    assert chisquare(off).pvalue > 1e-4
