@@ -314,6 +314,13 @@ __device__ __forceinline__ float2 fmul2(float2 a, float2 b) {
     return r;
 }
 
+// min(a, b, c) in one instruction (sm_100 family three-input min)
+__device__ __forceinline__ float fmin3(float a, float b, float c) {
+    float r;
+    asm("min.f32 %0, %1, %2, %3;" : "=f"(r) : "f"(a), "f"(b), "f"(c));
+    return r;
+}
+
 // v[i] for a lane-dependent i in [0, 32): binary select tree (no local memory).
 __device__ __forceinline__ uint32_t pick32(const uint32_t (&v)[32], int i) {
     uint32_t w16[16], w8[8], w4[4], w2[2];
@@ -393,6 +400,16 @@ __device__ __forceinline__ void screen_insert(ScreenRow &s, float L, int j) {
         return;
     }
     s.lev = fminf(s.lev, s.L[3]);
+    if (L < s.L[0] || (L == s.L[0] && j < s.J[0])) {  // a new head: shift the list down
+#pragma unroll
+        for (int t = TCAND - 1; t > 0; --t) {
+            s.L[t] = s.L[t - 1];
+            s.J[t] = s.J[t - 1];
+        }
+        s.L[0] = L;
+        s.J[0] = j;
+        return;
+    }
     float cl = L;
     int cj = j;
 #pragma unroll
@@ -799,13 +816,19 @@ __global__ void __launch_bounds__(tc_threads<NH>(), 1)
                         for (int g = 0; g < G; ++g) {
                             cm[g] = INFINITY;
 #pragma unroll
-                            for (int i = 8 * g; i < 8 * g + 8; i += 2) {
-                                const float2 c2 = reinterpret_cast<const float2 *>(rbuf)[(cc + i) >> 1];
-                                const float2 acc = make_float2(__uint_as_float(v[i]), __uint_as_float(v[i + 1]));
-                                const float2 st = ffma2(make_float2(-2.0f, -2.0f), acc, c2);
-                                cm[g] = fminf(cm[g], fminf(st.x, st.y));
-                                v[i] = __float_as_uint(st.x);
-                                v[i + 1] = __float_as_uint(st.y);
+                            for (int i = 8 * g; i < 8 * g + 8; i += 4) {
+                                // ||c||^2 of four columns in one 16-byte broadcast load
+                                const float4 c4 = reinterpret_cast<const float4 *>(rbuf)[(cc + i) >> 2];
+                                const float2 a0 = make_float2(__uint_as_float(v[i]), __uint_as_float(v[i + 1]));
+                                const float2 a1 = make_float2(__uint_as_float(v[i + 2]), __uint_as_float(v[i + 3]));
+                                const float2 s0 = ffma2(make_float2(-2.0f, -2.0f), a0, make_float2(c4.x, c4.y));
+                                const float2 s1 = ffma2(make_float2(-2.0f, -2.0f), a1, make_float2(c4.z, c4.w));
+                                cm[g] = fmin3(cm[g], s0.x, s0.y);
+                                cm[g] = fmin3(cm[g], s1.x, s1.y);
+                                v[i] = __float_as_uint(s0.x);
+                                v[i + 1] = __float_as_uint(s0.y);
+                                v[i + 2] = __float_as_uint(s1.x);
+                                v[i + 3] = __float_as_uint(s1.y);
                             }
                         }
                         if (SEG && (j0 < cb || j0 + SCR_CW > ce)) {
@@ -841,10 +864,16 @@ __global__ void __launch_bounds__(tc_threads<NH>(), 1)
                                         mask |= (__uint_as_float(v[i]) <= thr ? 1u : 0u) << i;
                                 }
                             }
-                            while (mask) {
-                                const int i = __ffs(mask) - 1;
-                                mask &= mask - 1;
-                                screen_insert(sr, __uint_as_float(pickn<SCR_CW>(v, i)), j0 + i);
+                            if ((mask & (mask - 1u)) == 0u) {
+                                // one column within the threshold (the usual case: a new
+                                // running minimum): it is the chunk's minimum
+                                screen_insert(sr, cmin, j0 + __ffs(mask) - 1);
+                            } else {
+                                while (mask) {
+                                    const int i = __ffs(mask) - 1;
+                                    mask &= mask - 1;
+                                    screen_insert(sr, __uint_as_float(pickn<SCR_CW>(v, i)), j0 + i);
+                                }
                             }
                         }
                     };
