@@ -231,8 +231,9 @@ def cpu_baseline_c4(Yb_host, C_host, K, budget_s=15.0):
         oracle.update_bf16(Yb_host[:ns], a, C_host)
         return time.perf_counter() - t0
 
-    t0 = one(200)
-    ns = int(min(Yb_host.shape[0], max(200, 200 * budget_s / max(t0, 1e-3))))
+    one(200)  # thread pool start-up
+    t0 = one(2000)
+    ns = int(min(Yb_host.shape[0], max(2000, 2000 * budget_s / max(t0, 1e-3))))
     t = one(ns)
     return ns * K / t, ns, t, oracle.num_threads()
 
