@@ -119,7 +119,14 @@ typedef struct skm_stats {
     int64_t prune_first_block;/* SKM_FLAG_PRUNE: (row, centroid) pairs alive
                                  after the first 32-dimension block             */
     int64_t prune_complete;   /* ... alive after the last block                 */
-    int64_t reserved[3];
+    double cluster_size_std;  /* population standard deviation of the k
+                                 cluster sizes of the final assignment (the
+                                 balance measure of the paper's Table 3)       */
+    int64_t *empty_per_iter;  /* INPUT: host int64 array of min(iters, 4096)
+                                 entries, or NULL; skm_fit writes the number of
+                                 empty clusters after each update (before any
+                                 split) of its first 4096 iterations           */
+    int64_t reserved;
 } skm_stats;
 
 const char *skm_last_error(void);
@@ -248,8 +255,10 @@ int skm_pca_fit(const float *X, int64_t n, int d, int d_out, float *mean, float 
  *    s_i = (max - b_i) / 255 (s_i = 1 for a flat dimension) when fit != 0,
  *    else the supplied b, s are used; code = clip(round((x - b)/s), 0, 255)
  *    in fp32, rounding half to even.  Outputs: codes uint8[n][d], b,s [d].
- *  repr = SKM_REPR_RBQ1 (RabitQ, 1-bit): mean m (fp64 sum, rounded to fp32)
- *    when fit != 0, else the supplied m; r = x - m; bit i = (r_i > 0);
+ *  repr = SKM_REPR_RBQ1 (RabitQ, 1-bit): mean m when fit != 0 (in exact
+ *    fixed point, see skm_mean_from_sums: m_c = fl32(S_c / (n 2^s)) with
+ *    S_c = sum of rint(x 2^s), s = skm_mean_scale(max |x|, n)), else the
+ *    supplied m; r = x - m; bit i = (r_i > 0);
  *    nx2 = ||r||^2; F = sqrt(d) ||r||^2 / ||r||_1 (0 when r = 0), i.e.
  *    ||r|| / <xbar, x>; popx = set bits.  nx2 and F come from compensated
  *    fp32 sums: within about 5 x 2^-24 and 12 x 2^-24 relative of the exact
@@ -284,6 +293,27 @@ typedef struct skm_quant_params {
 
 int skm_quantize(int repr, const float *X, int64_t n, int d, skm_quant_params *qp,
                  void *codes, void *ws, size_t ws_bytes, void *stream);
+
+/* The RabitQ dataset mean over row shards (one process per GPU), equal bit
+ * for bit to the single-process mean of skm_quantize(SKM_REPR_RBQ1, fit):
+ *  1. skm_column_absmax on each shard (device X float32 [n][d]; ws: device,
+ *     >= 4 bytes; writes max |x| to *amax_host; synchronises); take the
+ *     maximum over the shards;
+ *  2. s = skm_mean_scale(global max, total rows) (host): with 2^(E-1) <=
+ *     max |x| < 2^E and L = ceil(log2 n), s = 61 - L - E (0 when max = 0);
+ *  3. skm_column_sums_fixed on each shard ADDS sums[c] += S_c, the sum over
+ *     its rows of rint(x_rc 2^s) (round half to even; device int64 [d],
+ *     zeroed by the caller); every term is below 2^(61-L) in magnitude, so the sums are
+ *     exact integers and their order does not matter; sum S over the shards;
+ *  4. skm_mean_from_sums: m_c = fl32(fl64(S_c) / (n 2^s)) (one fp64
+ *     division, device float32 [d]).
+ * The fixed point keeps |m - mean| below 2^-(s+1) (about 2^-38 for unit-norm
+ * data and n = 10M).  Points must be finite.  Steps 3-4 are asynchronous. */
+int skm_column_absmax(const float *X, int64_t n, int d, float *amax_host, void *ws, size_t ws_bytes,
+                      void *stream);
+int skm_mean_scale(float amax, int64_t n_total);
+int skm_column_sums_fixed(const float *X, int64_t n, int d, int s, int64_t *sums, void *stream);
+int skm_mean_from_sums(const int64_t *sums, int64_t n_total, int d, int s, float *m, void *stream);
 
 /* Fixed-point exponent e of the RBQ1 decode-average: e = 24 - ceil(log2 max F)
  * (0 when every F is 0), so round(F 2^e) <= 2^24 (the largest F keeps its

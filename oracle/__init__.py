@@ -94,6 +94,9 @@ def lib():
                 "or_lvq4_exponent": ([vp, i64], i32),
                 "or_lvq4_update": ([vp, vp, i64, i32, i32, vp, i32, vp, vp], None),
                 "or_philox4x32_10": ([vp, vp, vp], None),
+                "or_mean_scale": ([ctypes.c_float, i64], i32),
+                "or_column_sums_fixed": ([vp, i64, i32, i32, vp], None),
+                "or_mean_from_sums": ([vp, i64, i32, i32, vp], None),
                 "or_forgy_indices": ([ctypes.c_uint64, i64, i32, vp], None),
             }
             for name, (args, res) in sig.items():
@@ -255,6 +258,28 @@ def rbq1_mean(X):
     n, d = X.shape
     m = np.empty(d, np.float32)
     lib().or_rbq1_mean(_p(X), n, d, _p(m))
+    return m
+
+
+def mean_scale(amax, n) -> int:
+    """Fixed-point scale s of the RabitQ mean for a maximum |x| and n rows."""
+    return int(lib().or_mean_scale(float(amax), int(n)))
+
+
+def column_sums_fixed(X, s):
+    """int64[d]: per column, the sum of rint(x 2^s) (exact)."""
+    X = _c(X, np.float32)
+    n, d = X.shape
+    S = np.zeros(d, np.int64)
+    lib().or_column_sums_fixed(_p(X), n, d, int(s), _p(S))
+    return S
+
+
+def mean_from_sums(S, n, s):
+    """fl32(fl64(S) / (n 2^s)) per column."""
+    S = _c(S, np.int64)
+    m = np.empty(S.shape[0], np.float32)
+    lib().or_mean_from_sums(_p(S), int(n), S.shape[0], int(s), _p(m))
     return m
 
 

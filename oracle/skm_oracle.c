@@ -310,12 +310,44 @@ double or_objective_bf16(const uint16_t *Xb, int64_t n, int d, const float *C,
 /* ------------------------------------------------------------------------ */
 
 /* Dataset mean m (fp64 sum, rounded to fp32). */
-void or_rbq1_mean(const float *X, int64_t n, int d, float *m) {
+/* The dataset mean m of Section 3.1 "RabitQ" in exact fixed point (the      */
+/* paper fixes no arithmetic for it): with 2^(E-1) <= max |x| < 2^E over all  */
+/* coordinates (frexp) and L = ceil(log2 n), s = 61 - L - E (0 when every x   */
+/* is 0); S_c = sum over the rows of rint(x_rc 2^s) as exact int64 (each      */
+/* term below 2^(61-L) in magnitude); m_c = fl32(fl64(S_c) / (n 2^s)).  Row   */
+/* shards summed at the same s give the same S_c.                            */
+/* Parity: pinned against the fp64 mean (|m - mean| <= 2^-(s+1) + half an    */
+/* fp32 ulp), exact means of grid data, and the shard sums.                  */
+int or_mean_scale(float amax, int64_t n) {
+    if (!(amax > 0.0f)) return 0;
+    int E = 0;
+    (void)frexpf(amax, &E); /* amax = f 2^E, f in [0.5, 1) */
+    int L = 0;
+    while (((int64_t)1 << L) < n) ++L;
+    return 61 - L - E;
+}
+
+void or_column_sums_fixed(const float *X, int64_t n, int d, int s, int64_t *S) {
     for (int i = 0; i < d; ++i) {
-        double s = 0.0;
-        for (int64_t p = 0; p < n; ++p) s += (double)X[p * (int64_t)d + i];
-        m[i] = (float)(s / (double)n);
+        int64_t acc = 0;
+        for (int64_t p = 0; p < n; ++p) acc += (int64_t)rint(ldexp((double)X[p * (int64_t)d + i], s));
+        S[i] += acc;
     }
+}
+
+void or_mean_from_sums(const int64_t *S, int64_t n, int d, int s, float *m) {
+    const double den = ldexp((double)n, s);
+    for (int i = 0; i < d; ++i) m[i] = (float)((double)S[i] / den);
+}
+
+void or_rbq1_mean(const float *X, int64_t n, int d, float *m) {
+    float amax = 0.0f;
+    for (int64_t t = 0; t < n * (int64_t)d; ++t) amax = fmaxf(amax, fabsf(X[t]));
+    const int s = or_mean_scale(amax, n);
+    int64_t *S = (int64_t *)calloc((size_t)d, sizeof(int64_t));
+    or_column_sums_fixed(X, n, d, s, S);
+    or_mean_from_sums(S, n, d, s, m);
+    free(S);
 }
 
 /* Per point: r = x - m (fp32); bit i = (r_i > 0), packed little-endian into

@@ -42,7 +42,8 @@ EXPORTED_SYMBOLS = [
     "skm_update",
     "skm_merge_partials", "skm_update_finalize", "skm_fit", "skm_split_empty", "skm_hier_workspace_size",
     "skm_fit_hierarchical", "skm_objective", "skm_sq8_decode", "skm_step_host_workspace_size",
-    "skm_lloyd_step_host", "skm_inject_fault", "skm_fault_armed", "skm_forgy_indices",
+    "skm_lloyd_step_host", "skm_inject_fault", "skm_fault_armed", "skm_forgy_indices", "skm_column_absmax",
+    "skm_mean_scale", "skm_column_sums_fixed", "skm_mean_from_sums",
 ]
 
 
@@ -74,7 +75,8 @@ class QuantParams(ctypes.Structure):
 class Stats(ctypes.Structure):
     _fields_ = [("rescored_rows", ctypes.c_int64), ("fallback_rows", ctypes.c_int64),
                 ("empty_clusters", ctypes.c_int64), ("prune_first_block", ctypes.c_int64),
-                ("prune_complete", ctypes.c_int64), ("reserved", ctypes.c_int64 * 3)]
+                ("prune_complete", ctypes.c_int64), ("cluster_size_std", ctypes.c_double),
+                ("empty_per_iter", ctypes.c_void_p), ("reserved", ctypes.c_int64)]
 
 
 class HierConfig(ctypes.Structure):
@@ -140,6 +142,10 @@ def lib():
             "skm_objective": ([vp, i32, i64, i32, vp, i32, vp, vp, vp, sz, vp], i32),
             "skm_sq8_decode": ([vp, i64, i32, vp, vp, vp, vp], i32),
             "skm_inject_fault": ([i32, i32], i32),
+            "skm_column_absmax": ([vp, i64, i32, vp, vp, sz, vp], i32),
+            "skm_mean_scale": ([ctypes.c_float, i64], i32),
+            "skm_column_sums_fixed": ([vp, i64, i32, i32, vp, vp], i32),
+            "skm_mean_from_sums": ([vp, i64, i32, i32, vp, vp], i32),
             "skm_fault_armed": ([i32], i32),
             "skm_step_host_workspace_size": ([vp, vp], sz),
             "skm_lloyd_step_host": ([vp, vp, vp, vp, vp, vp, vp, vp, sz, vp], i32),
@@ -475,12 +481,15 @@ def skm_fit(pts: Points, k, iters, C_init=None, init_idx=None, want_objective=Tr
     dist = torch.empty(pts.n, device=dev, dtype=torch.float32) if want_dist else None
     obj = (ctypes.c_double * (iters + 1))() if want_objective else None
     st = Stats()
+    empties = (ctypes.c_int64 * max(1, min(iters, 4096)))()
+    st.empty_per_iter = ctypes.cast(empties, ctypes.c_void_p)
     cfg = FitConfig(int(k), int(iters), int(empty_policy), 0, int(seed) & (2**64 - 1))
     _check(lib().skm_fit(ctypes.byref(cfg), ctypes.byref(pts.ref), _ptr(C_init), _ptr(init_idx), _ptr(C),
                          _ptr(assign), _ptr(dist), obj, ctypes.byref(st), _ptr(ws), ws.numel(), _stream(stream)))
     stats = {"rescored_rows": st.rescored_rows, "fallback_rows": st.fallback_rows,
              "empty_clusters": st.empty_clusters, "prune_first_block": st.prune_first_block,
-             "prune_complete": st.prune_complete}
+             "prune_complete": st.prune_complete, "cluster_size_std": st.cluster_size_std,
+             "empty_per_iter": list(empties)[:min(iters, 4096)]}
     return C, assign, dist, (list(obj) if obj is not None else None), stats
 
 
@@ -594,3 +603,29 @@ def skm_inject_fault(kind, count=1):
 
 def skm_fault_armed(kind) -> int:
     return int(lib().skm_fault_armed(int(kind)))
+
+
+def skm_column_absmax(X, stream=None) -> float:
+    """max |x| over a device float32 [n, d] tensor (synchronises)."""
+    n, d = X.shape
+    ws = _ws(256, X.device)
+    out = ctypes.c_float(0.0)
+    _check(lib().skm_column_absmax(_ptr(X), n, d, ctypes.byref(out), _ptr(ws), ws.numel(), _stream(stream)))
+    return float(out.value)
+
+
+def skm_mean_scale(amax, n_total) -> int:
+    return int(lib().skm_mean_scale(float(amax), int(n_total)))
+
+
+def skm_column_sums_fixed(X, s, sums, stream=None):
+    """sums (device int64 [d]) += per column, the sum of rint(x 2^s) over X's rows."""
+    n, d = X.shape
+    _check(lib().skm_column_sums_fixed(_ptr(X), n, d, int(s), _ptr(sums), _stream(stream)))
+    return sums
+
+
+def skm_mean_from_sums(sums, n_total, s, stream=None):
+    m = torch.empty(sums.numel(), device=sums.device, dtype=torch.float32)
+    _check(lib().skm_mean_from_sums(_ptr(sums), int(n_total), sums.numel(), int(s), _ptr(m), _stream(stream)))
+    return m

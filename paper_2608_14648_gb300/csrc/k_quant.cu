@@ -2,6 +2,8 @@
 // SQ8 and RabitQ 1-bit codes.  All kernels stream the fp32 points once with
 // 128-bit loads where the row length allows it; every float step that decides
 // a code is an explicit IEEE fp32 operation (no contraction).
+#include <string.h>
+
 #include "skm_internal.cuh"
 
 namespace skm {
@@ -461,6 +463,155 @@ __global__ void colmean_finish_kernel(const double *__restrict__ psum, int nblk,
     const double mu = __ddiv_rn(acc, (double)n);
     if (m) m[c] = __double2float_rn(mu);
     if (mean_d) mean_d[c] = mu;
+}
+
+// ---------------------------------------------------------------------------
+// The RabitQ dataset mean in exact fixed point: with 2^(E-1) <= max |x| < 2^E
+// over all points and L = ceil(log2 n), s = 61 - L - E; every coordinate
+// enters as rint(x 2^s) (an integer below 2^(61-L) in magnitude, formed from
+// the fp32 significand by fixed_rint), the column sums are exact int64 sums
+// (at most 2^61 in magnitude, order-independent), and m = fl32(S / (n 2^s))
+// with one fp64 division.  Row shards that use the same s and n add up to
+// exactly the single-process sums.
+// ---------------------------------------------------------------------------
+__host__ __device__ inline int mean_scale_of(unsigned amax_bits, int64_t n) {
+    if (amax_bits == 0) return 0;
+    const unsigned ef = (amax_bits >> 23) & 0xffu;
+    int E;
+    if (ef == 0) {  // subnormal maximum: mantissa m 2^-149, m < 2^23
+        unsigned mm = amax_bits & 0x7fffffu;
+        int hb = 0;
+        while (mm >> (hb + 1)) ++hb;
+        E = hb + 1 - 149;
+    } else {
+        E = (int)ef - 127 + 1;
+    }
+    int lg = 0;
+    while ((int64_t(1) << lg) < n) ++lg;
+    return 61 - lg - E;
+}
+
+__global__ void absmax_bits_kernel(const float *__restrict__ X, int64_t count, unsigned *__restrict__ bits) {
+    unsigned mx = 0;
+    const int64_t t0 = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
+    const int64_t st = (int64_t)gridDim.x * blockDim.x;
+    if (((uintptr_t)X & 15) == 0) {
+        const int64_t c4 = count >> 2;
+        const uint4 *X4 = reinterpret_cast<const uint4 *>(X);
+        for (int64_t i = t0; i < c4; i += st) {
+            const uint4 v = __ldg(X4 + i);
+            mx = max(mx, max(max(v.x & 0x7fffffffu, v.y & 0x7fffffffu), max(v.z & 0x7fffffffu, v.w & 0x7fffffffu)));
+        }
+        for (int64_t i = 4 * c4 + t0; i < count; i += st) mx = max(mx, __float_as_uint(X[i]) & 0x7fffffffu);
+    } else {
+        for (int64_t i = t0; i < count; i += st) mx = max(mx, __float_as_uint(X[i]) & 0x7fffffffu);
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) mx = max(mx, __shfl_xor_sync(0xffffffffu, mx, o));
+    if ((threadIdx.x & 31) == 0 && mx) atomicMax(bits, mx);
+}
+
+__global__ void mean_scale_kernel(const unsigned *__restrict__ bits, int64_t n, int *__restrict__ s_out) {
+    *s_out = mean_scale_of(*bits, n);
+}
+
+// S[c] += sum over this launch's rows of rint(x_rc 2^s); blocks take row
+// ranges, threads columns (four at a time when rows are 16-byte aligned).
+__global__ void colsum_fixed_kernel(const float *__restrict__ X, int64_t n, int d, const int *__restrict__ s_dev,
+                                    int s_host, unsigned long long *__restrict__ S) {
+    const int s = s_dev ? *s_dev : s_host;
+    const int64_t per = (n + gridDim.x - 1) / gridDim.x;
+    const int64_t r0 = (int64_t)blockIdx.x * per, r1 = min(n, r0 + per);
+    if (r0 >= r1) return;
+    if ((d & 3) == 0 && ((uintptr_t)X & 15) == 0) {
+        const int d4 = d >> 2;
+        const float4 *X4 = reinterpret_cast<const float4 *>(X);
+        for (int g = threadIdx.x; g < d4; g += blockDim.x) {
+            int64_t a0 = 0, a1 = 0, a2 = 0, a3 = 0;
+            int64_t r = r0;
+            for (; r + 4 <= r1; r += 4) {
+                float4 v[4];
+#pragma unroll
+                for (int u = 0; u < 4; ++u) v[u] = __ldg(X4 + (r + u) * d4 + g);
+#pragma unroll
+                for (int u = 0; u < 4; ++u) {
+                    a0 += fixed_rint(v[u].x, s);
+                    a1 += fixed_rint(v[u].y, s);
+                    a2 += fixed_rint(v[u].z, s);
+                    a3 += fixed_rint(v[u].w, s);
+                }
+            }
+            for (; r < r1; ++r) {
+                const float4 v = __ldg(X4 + r * d4 + g);
+                a0 += fixed_rint(v.x, s);
+                a1 += fixed_rint(v.y, s);
+                a2 += fixed_rint(v.z, s);
+                a3 += fixed_rint(v.w, s);
+            }
+            atomicAdd(S + 4 * g, (unsigned long long)a0);
+            atomicAdd(S + 4 * g + 1, (unsigned long long)a1);
+            atomicAdd(S + 4 * g + 2, (unsigned long long)a2);
+            atomicAdd(S + 4 * g + 3, (unsigned long long)a3);
+        }
+    } else {
+        for (int c = threadIdx.x; c < d; c += blockDim.x) {
+            int64_t a = 0;
+            for (int64_t r = r0; r < r1; ++r) a += fixed_rint(__ldg(X + r * d + c), s);
+            atomicAdd(S + c, (unsigned long long)a);
+        }
+    }
+}
+
+__global__ void mean_fixed_finish_kernel(const unsigned long long *__restrict__ S, int d, int64_t n,
+                                         const int *__restrict__ s_dev, int s_host, float *__restrict__ m) {
+    const int c = blockIdx.x * blockDim.x + threadIdx.x;
+    if (c >= d) return;
+    const int s = s_dev ? *s_dev : s_host;
+    const double q = __ddiv_rn(__ll2double_rn((long long)S[c]), scalbn((double)n, s));
+    m[c] = __double2float_rn(q);
+}
+
+int host_mean_scale(float amax, int64_t n) {
+    uint32_t b;
+    memcpy(&b, &amax, sizeof(b));
+    return mean_scale_of(b & 0x7fffffffu, n);
+}
+
+cudaError_t launch_absmax_bits(const float *X, int64_t count, unsigned *bits, cudaStream_t st) {
+    cudaError_t e = cudaMemsetAsync(bits, 0, sizeof(unsigned), st);
+    if (e != cudaSuccess) return e;
+    int64_t blocks = (count / 4 + 255) / 256;
+    blocks = blocks < 1 ? 1 : (blocks > 152 * 8 ? 152 * 8 : blocks);
+    absmax_bits_kernel<<<(unsigned)blocks, 256, 0, st>>>(X, count, bits);
+    return launched();
+}
+
+cudaError_t launch_mean_fixed(const float *X, int64_t n, int d, unsigned *bits, int *s_dev, unsigned long long *S,
+                              float *m, cudaStream_t st) {
+    cudaError_t e = launch_absmax_bits(X, n * (int64_t)d, bits, st);
+    if (e != cudaSuccess) return e;
+    mean_scale_kernel<<<1, 1, 0, st>>>(bits, n, s_dev);
+    if ((e = launched()) != cudaSuccess) return e;
+    if ((e = launch_colsum_fixed(X, n, d, s_dev, 0, S, true, st)) != cudaSuccess) return e;
+    return launch_mean_fixed_finish(S, d, n, s_dev, 0, m, st);
+}
+
+cudaError_t launch_colsum_fixed(const float *X, int64_t n, int d, const int *s_dev, int s_host,
+                                unsigned long long *S, bool zero_first, cudaStream_t st) {
+    if (zero_first) {
+        const cudaError_t e = cudaMemsetAsync(S, 0, sizeof(unsigned long long) * (size_t)d, st);
+        if (e != cudaSuccess) return e;
+    }
+    int64_t blocks = (n + 1023) / 1024;
+    blocks = blocks < 1 ? 1 : (blocks > 152 * 8 ? 152 * 8 : blocks);
+    colsum_fixed_kernel<<<(unsigned)blocks, 256, 0, st>>>(X, n, d, s_dev, s_host, S);
+    return launched();
+}
+
+cudaError_t launch_mean_fixed_finish(const unsigned long long *S, int d, int64_t n, const int *s_dev, int s_host,
+                                     float *m, cudaStream_t st) {
+    mean_fixed_finish_kernel<<<(d + 127) / 128, 128, 0, st>>>(S, d, n, s_dev, s_host, m);
+    return launched();
 }
 
 cudaError_t launch_colmean_finish(const double *psum, int nblk, int d, int64_t n, float *m,

@@ -37,6 +37,28 @@ __global__ void histogram_kernel(const int32_t *__restrict__ assign, int64_t n, 
     }
 }
 
+// One block: the number of zero entries of counts[0..k) into *out.
+__global__ void count_zeros_kernel(const int64_t *__restrict__ counts, int k, int64_t *__restrict__ out) {
+    __shared__ int part[32];
+    int z = 0;
+    for (int j = threadIdx.x; j < k; j += blockDim.x) z += counts[j] == 0;
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) z += __shfl_xor_sync(0xffffffffu, z, o);
+    if ((threadIdx.x & 31) == 0) part[threadIdx.x >> 5] = z;
+    __syncthreads();
+    if (threadIdx.x < 32) {
+        z = threadIdx.x < (blockDim.x >> 5) ? part[threadIdx.x] : 0;
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) z += __shfl_xor_sync(0xffffffffu, z, o);
+        if (threadIdx.x == 0) *out = z;
+    }
+}
+
+cudaError_t launch_count_zeros(const int64_t *counts, int k, int64_t *out, cudaStream_t st) {
+    count_zeros_kernel<<<1, 1024, 0, st>>>(counts, k, out);
+    return launched();
+}
+
 cudaError_t launch_histogram(const int32_t *assign, int64_t n, int k, int32_t *counts32,
                              cudaStream_t st) {
     cudaError_t e = cudaMemsetAsync(counts32, 0, sizeof(int32_t) * (size_t)k, st);

@@ -65,6 +65,7 @@ constexpr int64_t MAX_N_RBQ1 = int64_t(1) << 24;
 constexpr int64_t MAX_N_LVQ4 = int64_t(1) << 26;
 constexpr int RED_BLOCKS = 304;
 constexpr int PRUNE_MAX_D = 1024;  // 2 x 152 SMs for column / objective reductions
+constexpr int EMPTY_LOG = 4096;    // iterations whose empty-cluster counts skm_fit records
 
 static int check_data(const skm_data *x, bool need_codes = true) {
     if (!x) return set_error(SKM_ERR_INVALID_ARG, "skm_data is NULL");
@@ -201,6 +202,7 @@ struct FitBufs {
     int *status = nullptr;
     int64_t *counts = nullptr;
     int64_t *init_idx = nullptr;
+    int64_t *empty_iter = nullptr;  // empty clusters after each update (first EMPTY_LOG iterations)
 };
 
 static void plan_fit(const skm_data *x, int k, Carver &cv, FitBufs &b) {
@@ -222,6 +224,7 @@ static void plan_fit(const skm_data *x, int k, Carver &cv, FitBufs &b) {
     b.status = cv.take<int>(1);
     b.counts = cv.take<int64_t>(k);
     b.init_idx = cv.take<int64_t>(k);  // seeded Forgy indices (host-drawn)
+    b.empty_iter = cv.take<int64_t>(EMPTY_LOG);
 }
 
 static int need_ws(const Carver &cv, size_t ws_bytes, void *ws) {
@@ -601,9 +604,11 @@ int skm_quantize(int repr, const float *X, int64_t n, int d, skm_quant_params *q
         if (!qp->m || !qp->nx2 || !qp->F || !qp->popx)
             return set_error(SKM_ERR_INVALID_ARG, "RBQ1 needs m, nx2, F and popx");
         if (qp->fit) {
+            unsigned *bits = cv.take<unsigned>(1);
+            int *s_dev = cv.take<int>(1);
             SKM_TRY(need_ws(cv, ws_bytes, ws));
-            SKM_CUDA_TRY(launch_colsum_partial(X, n, d, psum, nblk, st));
-            SKM_CUDA_TRY(launch_colmean_finish(psum, nblk, d, n, qp->m, nullptr, st));
+            SKM_CUDA_TRY(launch_mean_fixed(X, n, d, bits, s_dev, reinterpret_cast<unsigned long long *>(psum), qp->m,
+                                           st));
         }
         SKM_CUDA_TRY(launch_rbq1_encode(X, n, d, qp->m, static_cast<uint32_t *>(codes), qp->nx2,
                                         qp->F, qp->popx, st));
@@ -632,6 +637,39 @@ int skm_lvq4_exponent(const float *lvq, int64_t n, int *e_host, void *ws, size_t
     SKM_CUDA_TRY(launch_lvq4_exponent(reinterpret_cast<const float4 *>(lvq), n, mb, ed, st));
     SKM_CUDA_TRY(cudaMemcpyAsync(e_host, ed, sizeof(int), cudaMemcpyDeviceToHost, st));
     SKM_CUDA_TRY(cudaStreamSynchronize(st));
+    return SKM_OK;
+}
+
+int skm_column_absmax(const float *X, int64_t n, int d, float *amax_host, void *ws, size_t ws_bytes, void *stream) {
+    if (!X || !amax_host || !ws) return set_error(SKM_ERR_INVALID_ARG, "NULL pointer");
+    if (n < 1 || d < 1 || d > MAX_D) return set_error(SKM_ERR_INVALID_ARG, "bad shape n=%lld d=%d", (long long)n, d);
+    if (ws_bytes < sizeof(unsigned)) return set_error(SKM_ERR_NO_MEMORY, "workspace too small");
+    cudaStream_t st = S(stream);
+    unsigned *bits = static_cast<unsigned *>(ws);
+    SKM_CUDA_TRY(launch_absmax_bits(X, n * (int64_t)d, bits, st));
+    unsigned h = 0;
+    SKM_CUDA_TRY(cudaMemcpyAsync(&h, bits, sizeof(h), cudaMemcpyDeviceToHost, st));
+    SKM_CUDA_TRY(cudaStreamSynchronize(st));
+    memcpy(amax_host, &h, sizeof(h));
+    return SKM_OK;
+}
+
+int skm_mean_scale(float amax, int64_t n_total) { return host_mean_scale(amax, n_total < 1 ? 1 : n_total); }
+
+int skm_column_sums_fixed(const float *X, int64_t n, int d, int s, int64_t *sums, void *stream) {
+    if (!X || !sums) return set_error(SKM_ERR_INVALID_ARG, "NULL pointer");
+    if (n < 1 || d < 1 || d > MAX_D) return set_error(SKM_ERR_INVALID_ARG, "bad shape n=%lld d=%d", (long long)n, d);
+    SKM_CUDA_TRY(
+        launch_colsum_fixed(X, n, d, nullptr, s, reinterpret_cast<unsigned long long *>(sums), false, S(stream)));
+    return SKM_OK;
+}
+
+int skm_mean_from_sums(const int64_t *sums, int64_t n_total, int d, int s, float *m, void *stream) {
+    if (!sums || !m) return set_error(SKM_ERR_INVALID_ARG, "NULL pointer");
+    if (n_total < 1 || d < 1 || d > MAX_D)
+        return set_error(SKM_ERR_INVALID_ARG, "bad shape n=%lld d=%d", (long long)n_total, d);
+    SKM_CUDA_TRY(launch_mean_fixed_finish(reinterpret_cast<const unsigned long long *>(sums), d, n_total, nullptr, s,
+                                          m, S(stream)));
     return SKM_OK;
 }
 
@@ -948,7 +986,10 @@ int skm_fit_hierarchical(const skm_hier_config *cfg, const skm_data *x, const in
     int32_t uflag = 0;
     SKM_CUDA_TRY(cudaMemcpy(&uflag, b.u.flag, sizeof(uflag), cudaMemcpyDeviceToHost));
     if (uflag) return set_error(SKM_ERR_TIMEOUT, "an update pipeline wait exceeded its limit");
-    if (stats_host) *stats_host = local;
+    if (stats_host) {
+        local.empty_per_iter = stats_host->empty_per_iter;  // an input field, left as given
+        *stats_host = local;
+    }
     return SKM_OK;
 }
 
@@ -1103,6 +1144,8 @@ int skm_fit(const skm_fit_config *cfg, const skm_data *x, const void *C_init,
         }
         if (it == cfg->iters) break;
         SKM_TRY(do_update(&xd, assign, k, C_out, b.counts, nullptr, e, b.u, st));
+        if (stats_host && stats_host->empty_per_iter && it < EMPTY_LOG)
+            SKM_CUDA_TRY(launch_count_zeros(b.counts, k, b.empty_iter + it, st));
         if (cfg->empty_policy == SKM_EMPTY_SPLIT)
             SKM_CUDA_TRY(launch_split_empty(C_out, x->repr == SKM_REPR_SQ8 ? 1 : 4, b.counts, k, x->d,
                                             b.u.wsplit, st));
@@ -1125,6 +1168,8 @@ int skm_fit(const skm_fit_config *cfg, const skm_data *x, const void *C_init,
     local.prune_first_block = (int64_t)pr[0];
     local.prune_complete = (int64_t)pr[1];
     if (stats_host) {
+        int64_t *per_iter = stats_host->empty_per_iter;
+        local.empty_per_iter = per_iter;
         *stats_host = local;
         std::vector<int64_t> cnt(k);
         if (cfg->iters > 0) {
@@ -1132,6 +1177,19 @@ int skm_fit(const skm_fit_config *cfg, const skm_data *x, const void *C_init,
                                     cudaMemcpyDeviceToHost));
             for (int j = 0; j < k; ++j) stats_host->empty_clusters += cnt[j] == 0;
         }
+        if (per_iter && cfg->iters > 0)
+            SKM_CUDA_TRY(cudaMemcpy(per_iter, b.empty_iter, sizeof(int64_t) * (size_t)std::min(cfg->iters, EMPTY_LOG),
+                                    cudaMemcpyDeviceToHost));
+        // balance of the final assignment: the standard deviation of the sizes
+        SKM_CUDA_TRY(launch_histogram(assign, n, k, b.u.counts32, st));
+        std::vector<int32_t> sz(k);
+        SKM_CUDA_TRY(cudaMemcpyAsync(sz.data(), b.u.counts32, sizeof(int32_t) * (size_t)k, cudaMemcpyDeviceToHost, st));
+        SKM_CUDA_TRY(cudaStreamSynchronize(st));
+        double mean = 0.0, var = 0.0;
+        for (int j = 0; j < k; ++j) mean += sz[j];
+        mean /= k;
+        for (int j = 0; j < k; ++j) var += (sz[j] - mean) * (sz[j] - mean);
+        stats_host->cluster_size_std = std::sqrt(var / k);
     }
     return SKM_OK;
 }

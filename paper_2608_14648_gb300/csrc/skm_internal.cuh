@@ -145,6 +145,17 @@ cudaError_t launch_sq8_decode(const uint8_t *codes, int64_t n, int d, const floa
                               const float *s, float *Y, cudaStream_t st);
 cudaError_t launch_colsum_partial(const float *X, int64_t n, int d, double *psum, int nblk,
                                   cudaStream_t st);
+// the RabitQ mean in exact fixed point (see k_quant.cu): the scale s of a
+// maximum |x| and a point count, the max |x| bits, the column sums at scale s
+// (added into S; s from s_dev when non-NULL, else s_host), and m = S / (n 2^s)
+int host_mean_scale(float amax, int64_t n);
+cudaError_t launch_absmax_bits(const float *X, int64_t count, unsigned *bits, cudaStream_t st);
+cudaError_t launch_colsum_fixed(const float *X, int64_t n, int d, const int *s_dev, int s_host,
+                                unsigned long long *S, bool zero_first, cudaStream_t st);
+cudaError_t launch_mean_fixed_finish(const unsigned long long *S, int d, int64_t n, const int *s_dev, int s_host,
+                                     float *m, cudaStream_t st);
+cudaError_t launch_mean_fixed(const float *X, int64_t n, int d, unsigned *bits, int *s_dev, unsigned long long *S,
+                              float *m, cudaStream_t st);
 cudaError_t launch_colmean_finish(const double *psum, int nblk, int d, int64_t n, float *m,
                                   double *mean_d, cudaStream_t st);
 cudaError_t launch_rbq1_encode(const float *X, int64_t n, int d, const float *m, uint32_t *codes,
@@ -191,6 +202,8 @@ cudaError_t launch_assign_rbq1(const uint32_t *codes, const float *nx2, const fl
 // update
 cudaError_t launch_histogram(const int32_t *assign, int64_t n, int k, int32_t *counts32,
                              cudaStream_t st);
+// *out = number of j < k with counts[j] == 0
+cudaError_t launch_count_zeros(const int64_t *counts, int k, int64_t *out, cudaStream_t st);
 cudaError_t launch_scan_offsets(const int32_t *counts32, int k, int64_t *offsets,
                                 int64_t *counts64_out, int accumulate_counts, cudaStream_t st);
 cudaError_t launch_scatter(const int32_t *assign, int64_t n, int k, const int64_t *offsets,

@@ -30,13 +30,36 @@ def allreduce_partials(partial: torch.Tensor, counts: torch.Tensor) -> None:
     dist.all_reduce(counts, op=dist.ReduceOp.SUM)
 
 
-def global_mean(local_sum: torch.Tensor, local_n: int) -> torch.Tensor:
-    """Dataset mean from per-rank column sums (fp64) and row counts."""
-    s = local_sum.to(torch.float64).clone()
-    cnt = torch.tensor([float(local_n)], dtype=torch.float64, device=s.device)
-    dist.all_reduce(s, op=dist.ReduceOp.SUM)
+def global_mean_fixed(amax_local: float, n_local: int, column_sums, mean_from_sums, device):
+    """The RabitQ dataset mean over all ranks' rows, the same bits as one
+    process computing it over all rows: the maximum of the ranks' max |x|
+    and the total row count give the fixed-point scale s (skm_mean_scale);
+    each rank's exact int64 column sums at that scale (column_sums(s)) are
+    summed over the ranks; mean_from_sums(S, n_total, s) finishes.  The two
+    callables carry the arithmetic (libskm on the GPU)."""
+    import paper_2608_14648_gb300 as skm
+
+    mx = torch.tensor([float(amax_local)], dtype=torch.float32, device=device)
+    cnt = torch.tensor([int(n_local)], dtype=torch.int64, device=device)
+    dist.all_reduce(mx, op=dist.ReduceOp.MAX)
     dist.all_reduce(cnt, op=dist.ReduceOp.SUM)
-    return (s / cnt).to(torch.float32)
+    n_total = int(cnt.item())
+    s = skm.skm_mean_scale(float(mx.item()), n_total)
+    S = column_sums(s)
+    dist.all_reduce(S, op=dist.ReduceOp.SUM)
+    return mean_from_sums(S, n_total, s)
+
+
+def global_rbq1_mean(X: torch.Tensor) -> torch.Tensor:
+    """global_mean_fixed with libskm's kernels on this rank's rows X (device float32 [n, d])."""
+    import paper_2608_14648_gb300 as skm
+
+    def sums(s):
+        S = torch.zeros(X.shape[1], dtype=torch.int64, device=X.device)
+        return skm.skm_column_sums_fixed(X, s, S)
+
+    return global_mean_fixed(skm.skm_column_absmax(X), X.shape[0], sums,
+                             lambda S, n, s: skm.skm_mean_from_sums(S, n, s), X.device)
 
 
 def global_exponent(local_e: int, device) -> int:

@@ -1,8 +1,9 @@
 """Multi-rank host logic on CPU (gloo, world_size 2): row sharding, the
-all-reduce of the update's partial sums and counts, the global mean and the
-global fixed-point exponent give the single-process result.  The partial
-sums here are plain numpy per shard (the same quantities skm_update writes
-with `partial`)."""
+all-reduce of the update's partial sums and counts, the global RabitQ mean
+and the global fixed-point exponent give the single-process result.  The
+partial sums here are plain numpy per shard (the same quantities skm_update
+writes with `partial`); the mean protocol runs with the oracle's fixed-point
+arithmetic and must give the single-process mean bit for bit."""
 import os
 import socket
 
@@ -12,6 +13,7 @@ import torch
 import torch.distributed as dist
 import torch.multiprocessing as mp
 
+import oracle
 from paper_2608_14648_gb300 import dist as skd
 
 
@@ -42,7 +44,13 @@ def _worker(rank, world, port, q):
         S, c = _partials(X[lo:hi], a[lo:hi], k, d)
         St, ct = torch.from_numpy(S), torch.from_numpy(c)
         skd.allreduce_partials(St, ct)
-        mean = skd.global_mean(torch.from_numpy(X[lo:hi].astype(np.float64).sum(0)), hi - lo)
+        import oracle
+
+        Xs = X[lo:hi]
+        mean = skd.global_mean_fixed(float(np.abs(Xs).max()), hi - lo,
+                                     lambda sc: torch.from_numpy(oracle.column_sums_fixed(Xs, sc)),
+                                     lambda S, nt, sc: torch.from_numpy(oracle.mean_from_sums(S.numpy(), nt, sc)),
+                                     "cpu")
         e = skd.global_exponent(30 + rank, "cpu")
         q.put((rank, St.numpy(), ct.numpy(), mean.numpy(), e, lo, hi))
     finally:
@@ -78,6 +86,6 @@ def test_two_rank_merge_equals_single_process():
     for rank, St, ct, mean, e, lo, hi in out:
         np.testing.assert_allclose(St, S, rtol=1e-12, atol=1e-12)
         np.testing.assert_array_equal(ct, c)
-        np.testing.assert_allclose(mean, X.astype(np.float64).mean(0), rtol=1e-6, atol=1e-7)
+        np.testing.assert_array_equal(mean, oracle.rbq1_mean(X))  # the single-process bits
         assert e == 30
     assert sorted((lo, hi) for _, _, _, _, _, lo, hi in out) == [(0, 501), (501, 1001)]

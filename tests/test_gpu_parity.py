@@ -287,7 +287,7 @@ def test_encode_rbq1_vs_oracle(skm, n, d):
     r = skm.skm_quantize(skm.REPR_RBQ1, X.to(DEV))
     h = _rbq1_host(r)
     m = oracle.rbq1_mean(X.numpy())
-    np.testing.assert_allclose(h["m"], m, rtol=1e-6, atol=1e-7)
+    np.testing.assert_array_equal(h["m"], m)  # the fixed-point mean, bit for bit
     # codes from the GPU's own mean must match the oracle's encoder bit for bit
     codes, nx2, F, popx = oracle.rbq1_encode(X.numpy(), h["m"])
     np.testing.assert_array_equal(h["codes"], codes)
@@ -1052,3 +1052,65 @@ def test_fit_seeded_forgy_matches_oracle(skm):
     Co, ao = oracle.lloyd_sq8(codes, codes[idx], iters)
     np.testing.assert_array_equal(a.cpu().numpy(), ao)
     np.testing.assert_array_equal(C.cpu().numpy(), Co)
+
+
+def test_fit_balance_statistics(skm):
+    """skm_stats: the per-iteration empty-cluster counts and the cluster-size
+    standard deviation of the final assignment (the balance column of the
+    paper's Table 3) equal the ones of the oracle's SQ8 trajectory (bit-exact
+    assignments, so the counts are the same integers)."""
+    n, d, k, iters = 3000, 32, 200, 5
+    X = _points(n, d, seed=81, ncomp=12)
+    q = skm.skm_quantize(skm.REPR_SQ8, X.to(DEV))
+    codes = q["codes"].cpu().numpy()
+    idx = synth.forgy_indices(n, k, seed=81)
+    idx[1:20:2] = idx[0:20:2]  # ten duplicated initial centroids: the higher copies start empty
+    _, a, _, _, st = skm.skm_fit(skm.Points(skm.REPR_SQ8, q["codes"], d), k, iters, init_idx=idx.to(DEV))
+    Cc = codes[idx.numpy()].copy()
+    empties = []
+    for _ in range(iters):
+        ao, _ = oracle.assign_sq8(codes, Cc)
+        Cc, co = oracle.update_sq8(codes, ao, Cc)
+        empties.append(int((co == 0).sum()))
+    ao, _ = oracle.assign_sq8(codes, Cc)
+    np.testing.assert_array_equal(a.cpu().numpy(), ao)
+    assert st["empty_per_iter"] == empties and max(empties) > 0
+    assert st["empty_clusters"] == empties[-1]
+    sizes = np.bincount(ao, minlength=k).astype(np.float64)
+    assert math.isclose(st["cluster_size_std"], float(sizes.std()), rel_tol=1e-12)
+
+
+@pytest.mark.parametrize("d", [768, 33])
+def test_sharded_rbq1_mean_codes_and_update_match_single(skm, d):
+    """Three uneven row shards: the merged fixed-point mean (shard max |x|,
+    scale from the global max and total rows, shard int64 column sums added)
+    equals the single-process skm_quantize mean bit for bit, so the shards'
+    codes and the merged fused decode-average equal the single-process ones."""
+    n, k = 5003, 23
+    X = _points(n, d, seed=91).to(DEV)
+    whole = skm.skm_quantize(skm.REPR_RBQ1, X)
+    bounds = [0, 17, 2950, n]
+    shards = [X[lo:hi].contiguous() for lo, hi in zip(bounds[:-1], bounds[1:])]
+    amax = max(skm.skm_column_absmax(xs) for xs in shards)
+    s = skm.skm_mean_scale(amax, n)
+    S = torch.zeros(d, dtype=torch.int64, device=DEV)
+    for xs in shards:
+        skm.skm_column_sums_fixed(xs, s, S)
+    m = skm.skm_mean_from_sums(S, n, s)
+    assert torch.equal(m, whole["m"])
+    pw = skm.rbq1_points(whole, d)
+    C = X[:k].clone()
+    a, _ = skm.skm_assign(pw, C)
+    C_single, cnt_single = skm.skm_update(pw, a, C.clone())
+    total = torch.zeros(k, d + 1, dtype=torch.int64, device=DEV)
+    counts = torch.zeros(k, dtype=torch.int64, device=DEV)
+    for (lo, hi), xs in zip(zip(bounds[:-1], bounds[1:]), shards):
+        q = skm.skm_quantize(skm.REPR_RBQ1, xs, fit=False, m=m.clone())
+        assert torch.equal(q["codes"], whole["codes"][lo:hi])
+        assert torch.equal(q["F"], whole["F"][lo:hi]) and torch.equal(q["nx2"], whole["nx2"][lo:hi])
+        sp = skm.Points(skm.REPR_RBQ1, q["codes"], d, q["nx2"], q["F"], q["popx"], m, pw.rbq1_exp)
+        part = torch.zeros(k, d + 1, dtype=torch.int64, device=DEV)
+        skm.skm_update(sp, a[lo:hi].contiguous(), None, counts=counts, partial=part)
+        skm.skm_merge_partials(total, part)
+    C_merged = skm.skm_update_finalize(pw, total, counts, C.clone())
+    assert torch.equal(counts, cnt_single) and torch.equal(C_merged, C_single)

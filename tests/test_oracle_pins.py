@@ -934,3 +934,45 @@ def test_forgy_indices_are_uniform():
     pairs = np.bincount(first * n + second, minlength=n * n).reshape(n, n)
     off = pairs[~np.eye(n, dtype=bool)]
     assert chisquare(off).pvalue > 1e-4
+
+
+# ------------------------------------------ RabitQ dataset mean in fixed point
+def test_mean_scale_by_hand():
+    # 1.0 = 0.5 * 2^1 -> E = 1; n = 1 -> L = 0; s = 61 - 0 - 1
+    assert oracle.mean_scale(1.0, 1) == 60
+    assert oracle.mean_scale(0.75, 1024) == 61 - 10 - 0
+    assert oracle.mean_scale(0.75, 1025) == 61 - 11 - 0
+    assert oracle.mean_scale(0.0, 100) == 0
+    assert oracle.mean_scale(2.0 ** -140, 2) == 61 - 1 + 139  # 2^-140 = 0.5 * 2^-139
+
+
+def test_rbq1_mean_is_the_mean_within_the_fixed_point_bound():
+    r = _rng(57)
+    n, d = 1000, 13
+    X = (r.standard_normal((n, d)) * np.logspace(-3, 1, d)).astype(np.float32)
+    m = oracle.rbq1_mean(X)
+    s = oracle.mean_scale(float(np.abs(X).max()), n)
+    exact = X.astype(np.float64).mean(axis=0)
+    bound = 2.0 ** -(s + 1) + np.abs(exact) * 2.0 ** -24 + 1e-300
+    assert np.all(np.abs(m.astype(np.float64) - exact) <= bound)
+
+
+def test_rbq1_mean_of_grid_data_is_exact():
+    """Coordinates on a 2^-10 grid: the fixed-point sums are the exact sums,
+    so m is the fp64 mean (exact sum, one division) rounded to fp32."""
+    r = _rng(58)
+    X = (r.integers(-4000, 4000, (777, 11)) / 1024.0).astype(np.float32)
+    want = (X.astype(np.float64).sum(axis=0) / 777).astype(np.float32)
+    np.testing.assert_array_equal(oracle.rbq1_mean(X), want)
+
+
+def test_rbq1_mean_shard_sums_add_up():
+    """Uneven row shards summed at the global scale give the whole-data sums,
+    hence the single-process mean bit for bit."""
+    r = _rng(59)
+    X = r.standard_normal((1001, 17)).astype(np.float32)
+    s = oracle.mean_scale(float(np.abs(X).max()), 1001)
+    parts = [X[:13], X[13:600], X[600:]]
+    S = sum(oracle.column_sums_fixed(p, s) for p in parts)
+    np.testing.assert_array_equal(S, oracle.column_sums_fixed(X, s))
+    np.testing.assert_array_equal(oracle.mean_from_sums(S, 1001, s), oracle.rbq1_mean(X))
