@@ -95,6 +95,11 @@ def lib():
                 "or_lvq4_update": ([vp, vp, i64, i32, i32, vp, i32, vp, vp], None),
                 "or_philox4x32_10": ([vp, vp, vp], None),
                 "or_mean_scale": ([ctypes.c_float, i64], i32),
+                "or_rbq1_seg_bounds": ([i32, vp, vp], None),
+                "or_rbq1_seg_encode": ([vp, i64, i32, vp, i32, i32, vp, vp, vp], None),
+                "or_rbq1_seg_centroid": ([vp, i32, i32, vp, i32, i32, vp, vp, vp, vp, vp], None),
+                "or_rbq1_seg_assign": ([vp, vp, vp, vp, i64, i32, i32, i32, vp, vp, vp, vp, vp, i32, vp, vp, vp],
+                                       None),
                 "or_column_sums_fixed": ([vp, i64, i32, i32, vp], None),
                 "or_mean_from_sums": ([vp, i64, i32, i32, vp], None),
                 "or_forgy_indices": ([ctypes.c_uint64, i64, i32, vp], None),
@@ -731,3 +736,57 @@ def forgy_indices(seed, n, k):
     out = np.empty(int(k), np.int64)
     lib().or_forgy_indices(ctypes.c_uint64(int(seed) & (2**64 - 1)), int(n), int(k), _p(out))
     return out
+
+
+# --------------------------------------------------------------------------
+# SuperKMeans with RabitQ codes: segment estimates and checkpoint pruning
+# --------------------------------------------------------------------------
+def rbq1_seg_bounds(d):
+    a, b = ctypes.c_int(0), ctypes.c_int(0)
+    lib().or_rbq1_seg_bounds(int(d), ctypes.byref(a), ctypes.byref(b))
+    return a.value, b.value
+
+
+def rbq1_seg_encode(X, m, bounds=None):
+    """Per point and segment: (nx2 f32[n, 3], F f32[n, 3], popx int32[n, 3])."""
+    X = _c(X, np.float32)
+    n, d = X.shape
+    d1, d2 = bounds if bounds is not None else rbq1_seg_bounds(d)
+    nx2 = np.empty((n, 3), np.float32)
+    F = np.empty((n, 3), np.float32)
+    pc = np.empty((n, 3), np.int32)
+    lib().or_rbq1_seg_encode(_p(X), n, d, _p(_c(m, np.float32)), d1, d2, _p(nx2), _p(F), _p(pc))
+    return nx2, F, pc
+
+
+def rbq1_seg_centroid(C, m, bounds=None):
+    """(ybar uint8[k, d], b f32[k], s f32[k], sumy int32[k, 3], ny2 f32[k, 3])."""
+    C = _c(C, np.float32)
+    k, d = C.shape
+    d1, d2 = bounds if bounds is not None else rbq1_seg_bounds(d)
+    ybar = np.empty((k, d), np.uint8)
+    b = np.empty(k, np.float32)
+    s = np.empty(k, np.float32)
+    sumy = np.empty((k, 3), np.int32)
+    ny2 = np.empty((k, 3), np.float32)
+    lib().or_rbq1_seg_centroid(_p(C), k, d, _p(_c(m, np.float32)), d1, d2, _p(ybar), _p(b), _p(s), _p(sumy),
+                               _p(ny2))
+    return ybar, b, s, sumy, ny2
+
+
+def rbq1_seg_assign(codes, seg, d, prep, prev=None, bounds=None):
+    """Checkpoint-pruned assignment (seg = rbq1_seg_encode output, prep =
+    rbq1_seg_centroid output).  Returns (assign int32[n], D3 f32[n])."""
+    codes = _c(codes, np.uint32)
+    nx2, F, pc = (_c(v, t) for v, t in zip(seg, (np.float32, np.float32, np.int32)))
+    ybar, b, s, sumy, ny2 = prep
+    n = codes.shape[0]
+    k = ybar.shape[0]
+    d1, d2 = bounds if bounds is not None else rbq1_seg_bounds(d)
+    a = np.empty(n, np.int32)
+    est = np.empty(n, np.float32)
+    pv = _c(prev, np.int32) if prev is not None else None
+    lib().or_rbq1_seg_assign(_p(codes), _p(nx2), _p(F), _p(pc), n, d, d1, d2, _p(_c(ybar, np.uint8)),
+                             _p(_c(b, np.float32)), _p(_c(s, np.float32)), _p(_c(sumy, np.int32)),
+                             _p(_c(ny2, np.float32)), k, _p(pv), _p(a), _p(est))
+    return a, est

@@ -970,3 +970,133 @@ void or_forgy_indices(uint64_t seed, int64_t n, int k, int64_t *out) {
     }
     free(a);
 }
+
+/* ------------------------------------------------------------------------ */
+/* SuperKMeans with RabitQ codes (Section 3.1 "SuperKMeans": for RabitQ the  */
+/* L2 distance decomposes over dimension segments, ||x - y||^2 = sum over    */
+/* segments of ||x_t - y_t||^2, each segment estimated with its own          */
+/* factors; pruning checkpoints after 12.5% and 25% of d).                   */
+/* Segments: [0, d1), [d1, d2), [d2, d) with d1 = 32 max(1, floor((d + 128)  */
+/* / 256)) (d/8 rounded to whole 32-dimension words) and d2 = 2 d1.          */
+/* Per point and segment t, with r = x - m (the global mean): nx2_t =        */
+/* ||r_t||^2, F_t = sqrt(d_t) ||r_t||^2 / ||r_t||_1 (0 when r_t = 0), both   */
+/* fp64 left to right rounded once; popx_t = set bits of the segment.        */
+/* Parity: the segment factors against their definitions; with the whole of  */
+/* d as one segment the estimate is the plain RabitQ one; on data lying on   */
+/* both grids the segment estimates are the exact segment distances.         */
+/* ------------------------------------------------------------------------ */
+void or_rbq1_seg_bounds(int d, int *d1, int *d2) {
+    int w = (d + 128) / 256;
+    if (w < 1) w = 1;
+    *d1 = 32 * w;
+    *d2 = 2 * (*d1);
+}
+
+void or_rbq1_seg_encode(const float *X, int64_t n, int d, const float *m, int d1, int d2, float *nx2s,
+                        float *Fs, int32_t *popxs) {
+    const int lo[3] = {0, d1, d2}, hi[3] = {d1, d2, d};
+#pragma omp parallel for schedule(static)
+    for (int64_t p = 0; p < n; ++p) {
+        for (int t = 0; t < 3; ++t) {
+            double s2 = 0.0, s1 = 0.0;
+            int32_t pc = 0;
+            for (int i = lo[t]; i < hi[t]; ++i) {
+                float r = X[p * (int64_t)d + i] - m[i];
+                if (r > 0.0f) pc += 1;
+                s2 += (double)r * (double)r;
+                s1 += fabs((double)r);
+            }
+            nx2s[p * 3 + t] = (float)s2;
+            Fs[p * 3 + t] = (s1 > 0.0) ? (float)(sqrt((double)(hi[t] - lo[t])) * s2 / s1) : 0.0f;
+            popxs[p * 3 + t] = pc;
+        }
+    }
+}
+
+/* Per centroid: the SQ4 codes of or_rbq1_centroid_sq4 (over all d), and per  */
+/* segment the code sum and ||rho_t||^2 (the blocked fp64 order of           */
+/* sumsq_blocked over the segment's words).                                   */
+void or_rbq1_seg_centroid(const float *C, int k, int d, const float *m, int d1, int d2, uint8_t *ybar,
+                          float *b, float *s, int32_t *sumy3, float *ny2s) {
+    int32_t *sumy = (int32_t *)malloc(sizeof(int32_t) * (size_t)k);
+    float *ny2 = (float *)malloc(sizeof(float) * (size_t)k);
+    or_rbq1_centroid_sq4(C, k, d, m, ybar, b, s, sumy, ny2);
+    float *rho = (float *)malloc(sizeof(float) * (size_t)d);
+    const int lo[3] = {0, d1, d2}, hi[3] = {d1, d2, d};
+    for (int j = 0; j < k; ++j) {
+        for (int i = 0; i < d; ++i) rho[i] = C[(int64_t)j * d + i] - m[i];
+        for (int t = 0; t < 3; ++t) {
+            int32_t sy = 0;
+            for (int i = lo[t]; i < hi[t]; ++i) sy += ybar[(int64_t)j * d + i];
+            sumy3[(int64_t)j * 3 + t] = sy;
+            ny2s[(int64_t)j * 3 + t] = (float)sumsq_blocked(rho + lo[t], hi[t] - lo[t]);
+        }
+    }
+    free(rho);
+    free(sumy);
+    free(ny2);
+}
+
+/* Segment estimate of Eq. rabitq_l2 with Eq. final:rabitq on the segment, in  */
+/* the library's fp32 order: isd_t = fl(1/sqrt(d_t)), sd = s isd_t, bd = b    */
+/* isd_t, u = fma(sd, 2 P_t - sumy_t, bd (2 popx_t - d_t)), est = fma(-2 F_t,  */
+/* u, nx2_t + ny2_t).  Partial estimates D1 = est_0, D2 = D1 + est_1,         */
+/* D3 = D2 + est_2 (fp32).                                                    */
+/* Pruning (an order-independent reading of the checkpoints): the bound is    */
+/* beta = D3 of the row's seed centroid (its previous assignment, entries     */
+/* outside [0, k) and prev = NULL meaning centroid 0); a centroid other than  */
+/* the seed stays a candidate only if D1 <= beta and D2 <= beta; the result   */
+/* is the candidate (seed included) with the smallest D3, ties to the lowest  */
+/* index.  est_best receives that D3.                                         */
+void or_rbq1_seg_assign(const uint32_t *codes, const float *nx2s, const float *Fs, const int32_t *popxs,
+                        int64_t n, int d, int d1, int d2, const uint8_t *ybar, const float *b, const float *s,
+                        const int32_t *sumy3, const float *ny2s, int k, const int32_t *prev, int32_t *assign,
+                        float *est_best) {
+    const int W = (d + 31) / 32;
+    const int lo[3] = {0, d1, d2}, hi[3] = {d1, d2, d};
+    float isd[3];
+    for (int t = 0; t < 3; ++t) isd[t] = hi[t] > lo[t] ? (float)(1.0 / sqrt((double)(hi[t] - lo[t]))) : 0.0f;
+#pragma omp parallel for schedule(dynamic, 16)
+    for (int64_t p = 0; p < n; ++p) {
+        const uint32_t *cw = codes + p * (int64_t)W;
+        float D[3];
+        int seed = prev ? prev[p] : 0;
+        if (seed < 0 || seed >= k) seed = 0;
+        float beta = 0.0f;
+        for (int pass = 0; pass < 2; ++pass) {
+            float best = INFINITY;
+            int32_t a = -1;
+            for (int j = (pass == 0 ? seed : 0); j < (pass == 0 ? seed + 1 : k); ++j) {
+                const uint8_t *y = ybar + (int64_t)j * d;
+                int alive = 1;
+                for (int t = 0; t < 3 && alive; ++t) {
+                    if (hi[t] == lo[t]) { /* an empty segment adds nothing */
+                        D[t] = (t == 0) ? 0.0f : D[t - 1];
+                        continue;
+                    }
+                    int32_t P = 0;
+                    for (int i = lo[t]; i < hi[t]; ++i)
+                        if ((cw[i / 32] >> (i % 32)) & 1u) P += y[i];
+                    const float sd = s[j] * isd[t];
+                    const float bd = b[j] * isd[t];
+                    const float pc = (float)(2 * popxs[p * 3 + t] - (hi[t] - lo[t]));
+                    const float u = fmaf(sd, (float)(2 * P - sumy3[(int64_t)j * 3 + t]), bd * pc);
+                    const float est = fmaf(-2.0f * Fs[p * 3 + t], u, nx2s[p * 3 + t] + ny2s[(int64_t)j * 3 + t]);
+                    D[t] = (t == 0) ? est : D[t - 1] + est;
+                    if (pass == 1 && t < 2 && j != seed && !(D[t] <= beta)) alive = 0;
+                }
+                if (!alive) continue;
+                if (D[2] < best) {
+                    best = D[2];
+                    a = j;
+                }
+            }
+            if (pass == 0) {
+                beta = best;
+            } else {
+                assign[p] = a;
+                if (est_best) est_best[p] = best;
+            }
+        }
+    }
+}

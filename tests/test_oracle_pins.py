@@ -976,3 +976,79 @@ def test_rbq1_mean_shard_sums_add_up():
     S = sum(oracle.column_sums_fixed(p, s) for p in parts)
     np.testing.assert_array_equal(S, oracle.column_sums_fixed(X, s))
     np.testing.assert_array_equal(oracle.mean_from_sums(S, 1001, s), oracle.rbq1_mean(X))
+
+
+# ---------------------------------- SuperKMeans with RabitQ: segment estimates
+def test_rbq1_seg_bounds():
+    assert oracle.rbq1_seg_bounds(1024) == (128, 256)  # 12.5% and 25% of d
+    assert oracle.rbq1_seg_bounds(768) == (96, 192)
+    assert oracle.rbq1_seg_bounds(128) == (32, 64)
+
+
+def test_rbq1_seg_factors_are_their_definitions():
+    r = _rng(61)
+    n, d = 30, 256
+    X = r.standard_normal((n, d)).astype(np.float32)
+    m = oracle.rbq1_mean(X)
+    d1, d2 = oracle.rbq1_seg_bounds(d)
+    nx2, F, pc = oracle.rbq1_seg_encode(X, m)
+    R = X.astype(np.float64) - m.astype(np.float64)
+    for t, (lo, hi) in enumerate([(0, d1), (d1, d2), (d2, d)]):
+        Rt = R[:, lo:hi]
+        s2, s1 = (Rt ** 2).sum(1), np.abs(Rt).sum(1)
+        np.testing.assert_allclose(nx2[:, t], s2, rtol=1e-6)
+        np.testing.assert_allclose(F[:, t], math.sqrt(hi - lo) * s2 / s1, rtol=1e-6)
+        np.testing.assert_array_equal(pc[:, t], ((X[:, lo:hi] - m[lo:hi]) > 0).sum(1))
+
+
+def test_rbq1_seg_whole_d_is_plain_rabitq():
+    """One segment spanning all of d (the other two empty): the segment
+    estimate is the plain RabitQ estimate, and with the bound from centroid 0
+    the pruned argmin is the plain argmin."""
+    r = _rng(62)
+    n, d, k = 200, 96, 9
+    X = r.standard_normal((n, d)).astype(np.float32)
+    C = r.standard_normal((k, d)).astype(np.float32)
+    m = oracle.rbq1_mean(X)
+    codes, nx2, F, popx = oracle.rbq1_encode(X, m)
+    seg = oracle.rbq1_seg_encode(X, m, bounds=(d, d))
+    np.testing.assert_array_equal(seg[0][:, 0], nx2)
+    np.testing.assert_array_equal(seg[1][:, 0], F)
+    np.testing.assert_array_equal(seg[2][:, 0], popx)
+    a0, e0 = oracle.rbq1_assign(codes, nx2, F, popx, d, oracle.rbq1_centroid_sq4(C, m))
+    a1, e1 = oracle.rbq1_seg_assign(codes, seg, d, oracle.rbq1_seg_centroid(C, m, bounds=(d, d)), bounds=(d, d))
+    np.testing.assert_array_equal(a1, a0)
+    np.testing.assert_array_equal(e1, e0)
+
+
+def test_rbq1_seg_estimates_exact_on_grid_and_pruning_keeps_the_nearest():
+    """Residuals of constant magnitude within each segment (the 1-bit code
+    then reconstructs each segment exactly) and centroids on SQ4 grids: every
+    segment estimate is the exact segment distance, the partial estimates are
+    partial distances, and the checkpoint pruning returns the true nearest
+    centroid whatever the seed of its bound."""
+    r = _rng(63)
+    n, d, k = 60, 256, 8
+    d1, d2 = oracle.rbq1_seg_bounds(d)
+    m = np.zeros(d, np.float32)
+    amp = np.empty((n, d), np.float64)
+    for lo, hi in [(0, d1), (d1, d2), (d2, d)]:
+        amp[:, lo:hi] = r.uniform(0.25, 2.0, (n, 1))
+    X = (amp * np.where(r.random((n, d)) < 0.5, -1.0, 1.0)).astype(np.float32)
+    yb = r.integers(0, 16, (k, d))
+    yb[:, 0], yb[:, 1] = 0, 15
+    b0 = r.choice([-1.0, -0.75, -0.5], k).astype(np.float32)
+    s0 = r.choice([0.0625, 0.125, 0.25], k).astype(np.float32)
+    C = (b0[:, None] + s0[:, None] * yb).astype(np.float32)
+    seg = oracle.rbq1_seg_encode(X, m)
+    prep = oracle.rbq1_seg_centroid(C, m)
+    codes, _, _, _ = oracle.rbq1_encode(X, m)
+    true = cdist(X.astype(np.float64), C.astype(np.float64), "sqeuclidean")
+    want = np.argmin(true, axis=1)
+    gap = np.sort(true, axis=1)
+    assert np.all(gap[:, 1] - gap[:, 0] > 1e-3 * gap[:, 0])  # no near ties
+    for prev in (None, np.zeros(n, np.int32), np.full(n, k - 1, np.int32), want.astype(np.int32),
+                 r.integers(0, k, n).astype(np.int32)):
+        a, est = oracle.rbq1_seg_assign(codes, seg, d, prep, prev=prev)
+        np.testing.assert_array_equal(a, want)
+        np.testing.assert_allclose(est, true[np.arange(n), want], rtol=1e-5)
