@@ -98,8 +98,10 @@ def lib():
                 "or_rbq1_seg_bounds": ([i32, vp, vp], None),
                 "or_rbq1_seg_encode": ([vp, i64, i32, vp, i32, i32, vp, vp, vp], None),
                 "or_rbq1_seg_centroid": ([vp, i32, i32, vp, i32, i32, vp, vp, vp, vp, vp], None),
-                "or_rbq1_seg_assign": ([vp, vp, vp, vp, i64, i32, i32, i32, vp, vp, vp, vp, vp, i32, vp, vp, vp],
-                                       None),
+                "or_rbq1_seg_assign": ([vp, vp, vp, vp, i64, i32, i32, i32, vp, vp, vp, vp, vp, i32, vp, vp, vp,
+                                        vp], None),
+                "or_rbq1_seg_factors": ([i32, i32, i32, f64, vp], None),
+                "or_rbq1_seg_partials": ([vp, vp, vp, vp, i64, i32, i32, i32, vp, vp, vp, vp, vp, i32, vp], None),
                 "or_column_sums_fixed": ([vp, i64, i32, i32, vp], None),
                 "or_mean_from_sums": ([vp, i64, i32, i32, vp], None),
                 "or_forgy_indices": ([ctypes.c_uint64, i64, i32, vp], None),
@@ -774,9 +776,24 @@ def rbq1_seg_centroid(C, m, bounds=None):
     return ybar, b, s, sumy, ny2
 
 
-def rbq1_seg_assign(codes, seg, d, prep, prev=None, bounds=None):
+SEG_EPS0 = 2.1  # ADSampling's default significance parameter
+
+
+def rbq1_seg_factors(d, bounds=None, eps0=SEG_EPS0):
+    """Checkpoint factors g_t = fl32((e_t / d) (1 + eps0 / sqrt(e_t))^2)."""
+    d1, d2 = bounds if bounds is not None else rbq1_seg_bounds(d)
+    g = np.empty(2, np.float32)
+    lib().or_rbq1_seg_factors(int(d), d1, d2, float(eps0), _p(g))
+    return g
+
+
+def rbq1_seg_assign(codes, seg, d, prep, prev=None, bounds=None, g=None):
     """Checkpoint-pruned assignment (seg = rbq1_seg_encode output, prep =
-    rbq1_seg_centroid output).  Returns (assign int32[n], D3 f32[n])."""
+    rbq1_seg_centroid output, g = the two checkpoint factors, default
+    ADSampling's with eps0 = 2.1; g = (1, 1) is the exact test).  Returns
+    (assign int32[n], D3 f32[n])."""
+    if g is None:
+        g = rbq1_seg_factors(d, bounds)
     codes = _c(codes, np.uint32)
     nx2, F, pc = (_c(v, t) for v, t in zip(seg, (np.float32, np.float32, np.int32)))
     ybar, b, s, sumy, ny2 = prep
@@ -788,5 +805,19 @@ def rbq1_seg_assign(codes, seg, d, prep, prev=None, bounds=None):
     pv = _c(prev, np.int32) if prev is not None else None
     lib().or_rbq1_seg_assign(_p(codes), _p(nx2), _p(F), _p(pc), n, d, d1, d2, _p(_c(ybar, np.uint8)),
                              _p(_c(b, np.float32)), _p(_c(s, np.float32)), _p(_c(sumy, np.int32)),
-                             _p(_c(ny2, np.float32)), k, _p(pv), _p(a), _p(est))
+                             _p(_c(ny2, np.float32)), k, _p(pv), _p(_c(g, np.float32)), _p(a), _p(est))
     return a, est
+
+
+def rbq1_seg_partials(codes, seg, d, prep, bounds=None):
+    """Every pair's partial estimates (D1, D2, D3): f32[n, k, 3]."""
+    codes = _c(codes, np.uint32)
+    nx2, F, pc = (_c(v, t) for v, t in zip(seg, (np.float32, np.float32, np.int32)))
+    ybar, b, s, sumy, ny2 = prep
+    n, k = codes.shape[0], ybar.shape[0]
+    d1, d2 = bounds if bounds is not None else rbq1_seg_bounds(d)
+    D = np.empty((n, k, 3), np.float32)
+    lib().or_rbq1_seg_partials(_p(codes), _p(nx2), _p(F), _p(pc), n, d, d1, d2, _p(_c(ybar, np.uint8)),
+                               _p(_c(b, np.float32)), _p(_c(s, np.float32)), _p(_c(sumy, np.int32)),
+                               _p(_c(ny2, np.float32)), k, _p(D))
+    return D

@@ -1044,14 +1044,46 @@ void or_rbq1_seg_centroid(const float *C, int k, int d, const float *m, int d1, 
 /* D3 = D2 + est_2 (fp32).                                                    */
 /* Pruning (an order-independent reading of the checkpoints): the bound is    */
 /* beta = D3 of the row's seed centroid (its previous assignment, entries     */
-/* outside [0, k) and prev = NULL meaning centroid 0); a centroid other than  */
-/* the seed stays a candidate only if D1 <= beta and D2 <= beta; the result   */
-/* is the candidate (seed included) with the smallest D3, ties to the lowest  */
-/* index.  est_best receives that D3.                                         */
+/* outside [0, k) and prev = NULL meaning centroid 0); at checkpoint t (after */
+/* e_t = d1, d2 dimensions) a centroid other than the seed is dropped when    */
+/* D_t > fl32(beta g_t), g_t the checkpoint's factor: ADSampling's test       */
+/* D_t d / e_t > beta (1 + eps0 / sqrt(e_t))^2 gives g_t = fl32((e_t / d)     */
+/* (1 + eps0 / sqrt(e_t))^2) (or_rbq1_seg_factors, eps0 = 2.1), g_t = 1 the   */
+/* exact test; the result is the candidate (seed included) with the smallest  */
+/* D3, ties to the lowest index.  est_best receives that D3.                  */
+void or_rbq1_seg_factors(int d, int d1, int d2, double eps0, float *g) {
+    const int e[2] = {d1, d2};
+    for (int t = 0; t < 2; ++t) {
+        const double a = 1.0 + eps0 / sqrt((double)e[t]);
+        g[t] = (float)(((double)e[t] / (double)d) * a * a);
+    }
+}
+
+/* The partial estimates D1, D2, D3 of point p against centroid j. */
+static void seg_partials(const uint32_t *cw, const float *nx2s, const float *Fs, const int32_t *popxs, int64_t p,
+                         int d, const int lo[3], const int hi[3], const float isd[3], const uint8_t *y, float b,
+                         float s, const int32_t *sumy3, const float *ny2s, float D[3]) {
+    for (int t = 0; t < 3; ++t) {
+        if (hi[t] == lo[t]) { /* an empty segment adds nothing */
+            D[t] = (t == 0) ? 0.0f : D[t - 1];
+            continue;
+        }
+        int32_t P = 0;
+        for (int i = lo[t]; i < hi[t]; ++i)
+            if ((cw[i / 32] >> (i % 32)) & 1u) P += y[i];
+        const float sd = s * isd[t];
+        const float bd = b * isd[t];
+        const float pc = (float)(2 * popxs[p * 3 + t] - (hi[t] - lo[t]));
+        const float u = fmaf(sd, (float)(2 * P - sumy3[t]), bd * pc);
+        const float est = fmaf(-2.0f * Fs[p * 3 + t], u, nx2s[p * 3 + t] + ny2s[t]);
+        D[t] = (t == 0) ? est : D[t - 1] + est;
+    }
+}
+
 void or_rbq1_seg_assign(const uint32_t *codes, const float *nx2s, const float *Fs, const int32_t *popxs,
                         int64_t n, int d, int d1, int d2, const uint8_t *ybar, const float *b, const float *s,
-                        const int32_t *sumy3, const float *ny2s, int k, const int32_t *prev, int32_t *assign,
-                        float *est_best) {
+                        const int32_t *sumy3, const float *ny2s, int k, const int32_t *prev, const float *g,
+                        int32_t *assign, float *est_best) {
     const int W = (d + 31) / 32;
     const int lo[3] = {0, d1, d2}, hi[3] = {d1, d2, d};
     float isd[3];
@@ -1059,44 +1091,39 @@ void or_rbq1_seg_assign(const uint32_t *codes, const float *nx2s, const float *F
 #pragma omp parallel for schedule(dynamic, 16)
     for (int64_t p = 0; p < n; ++p) {
         const uint32_t *cw = codes + p * (int64_t)W;
-        float D[3];
         int seed = prev ? prev[p] : 0;
         if (seed < 0 || seed >= k) seed = 0;
-        float beta = 0.0f;
-        for (int pass = 0; pass < 2; ++pass) {
-            float best = INFINITY;
-            int32_t a = -1;
-            for (int j = (pass == 0 ? seed : 0); j < (pass == 0 ? seed + 1 : k); ++j) {
-                const uint8_t *y = ybar + (int64_t)j * d;
-                int alive = 1;
-                for (int t = 0; t < 3 && alive; ++t) {
-                    if (hi[t] == lo[t]) { /* an empty segment adds nothing */
-                        D[t] = (t == 0) ? 0.0f : D[t - 1];
-                        continue;
-                    }
-                    int32_t P = 0;
-                    for (int i = lo[t]; i < hi[t]; ++i)
-                        if ((cw[i / 32] >> (i % 32)) & 1u) P += y[i];
-                    const float sd = s[j] * isd[t];
-                    const float bd = b[j] * isd[t];
-                    const float pc = (float)(2 * popxs[p * 3 + t] - (hi[t] - lo[t]));
-                    const float u = fmaf(sd, (float)(2 * P - sumy3[(int64_t)j * 3 + t]), bd * pc);
-                    const float est = fmaf(-2.0f * Fs[p * 3 + t], u, nx2s[p * 3 + t] + ny2s[(int64_t)j * 3 + t]);
-                    D[t] = (t == 0) ? est : D[t - 1] + est;
-                    if (pass == 1 && t < 2 && j != seed && !(D[t] <= beta)) alive = 0;
-                }
-                if (!alive) continue;
-                if (D[2] < best) {
-                    best = D[2];
-                    a = j;
-                }
-            }
-            if (pass == 0) {
-                beta = best;
-            } else {
-                assign[p] = a;
-                if (est_best) est_best[p] = best;
+        float D[3];
+        seg_partials(cw, nx2s, Fs, popxs, p, d, lo, hi, isd, ybar + (int64_t)seed * d, b[seed], s[seed],
+                     sumy3 + (int64_t)seed * 3, ny2s + (int64_t)seed * 3, D);
+        const float beta = D[2];
+        float best = INFINITY;
+        int32_t a = -1;
+        for (int j = 0; j < k; ++j) {
+            seg_partials(cw, nx2s, Fs, popxs, p, d, lo, hi, isd, ybar + (int64_t)j * d, b[j], s[j],
+                         sumy3 + (int64_t)j * 3, ny2s + (int64_t)j * 3, D);
+            if (j != seed && (D[0] > beta * g[0] || D[1] > beta * g[1])) continue;
+            if (D[2] < best) {
+                best = D[2];
+                a = j;
             }
         }
+        assign[p] = a;
+        if (est_best) est_best[p] = best;
     }
+}
+
+/* Every pair's partial estimates D[p][j][0..2] (no pruning). */
+void or_rbq1_seg_partials(const uint32_t *codes, const float *nx2s, const float *Fs, const int32_t *popxs,
+                          int64_t n, int d, int d1, int d2, const uint8_t *ybar, const float *b, const float *s,
+                          const int32_t *sumy3, const float *ny2s, int k, float *D) {
+    const int W = (d + 31) / 32;
+    const int lo[3] = {0, d1, d2}, hi[3] = {d1, d2, d};
+    float isd[3];
+    for (int t = 0; t < 3; ++t) isd[t] = hi[t] > lo[t] ? (float)(1.0 / sqrt((double)(hi[t] - lo[t]))) : 0.0f;
+#pragma omp parallel for schedule(static)
+    for (int64_t p = 0; p < n; ++p)
+        for (int j = 0; j < k; ++j)
+            seg_partials(codes + p * (int64_t)W, nx2s, Fs, popxs, p, d, lo, hi, isd, ybar + (int64_t)j * d, b[j],
+                         s[j], sumy3 + (int64_t)j * 3, ny2s + (int64_t)j * 3, D + (p * (int64_t)k + j) * 3);
 }

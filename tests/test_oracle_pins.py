@@ -1025,8 +1025,8 @@ def test_rbq1_seg_estimates_exact_on_grid_and_pruning_keeps_the_nearest():
     """Residuals of constant magnitude within each segment (the 1-bit code
     then reconstructs each segment exactly) and centroids on SQ4 grids: every
     segment estimate is the exact segment distance, the partial estimates are
-    partial distances, and the checkpoint pruning returns the true nearest
-    centroid whatever the seed of its bound."""
+    partial distances, and the checkpoint pruning with the exact test (g = 1)
+    returns the true nearest centroid whatever the seed of its bound."""
     r = _rng(63)
     n, d, k = 60, 256, 8
     d1, d2 = oracle.rbq1_seg_bounds(d)
@@ -1049,6 +1049,39 @@ def test_rbq1_seg_estimates_exact_on_grid_and_pruning_keeps_the_nearest():
     assert np.all(gap[:, 1] - gap[:, 0] > 1e-3 * gap[:, 0])  # no near ties
     for prev in (None, np.zeros(n, np.int32), np.full(n, k - 1, np.int32), want.astype(np.int32),
                  r.integers(0, k, n).astype(np.int32)):
-        a, est = oracle.rbq1_seg_assign(codes, seg, d, prep, prev=prev)
+        a, est = oracle.rbq1_seg_assign(codes, seg, d, prep, prev=prev, g=np.ones(2, np.float32))
         np.testing.assert_array_equal(a, want)
         np.testing.assert_allclose(est, true[np.arange(n), want], rtol=1e-5)
+
+
+def test_rbq1_seg_pruning_rule_brute_force():
+    """The scaled checkpoint test (ADSampling's factors) against the rule
+    restated over every pair's partial estimates: the candidates are the seed
+    and every centroid whose partial estimates stay <= fl32(beta g_t), the
+    result the candidate with the smallest D3 (lowest index on ties)."""
+    r = _rng(64)
+    n, d, k = 50, 256, 40
+    X = r.standard_normal((n, d)).astype(np.float32)
+    C = (X[r.integers(0, n, k)] + 0.3 * r.standard_normal((k, d))).astype(np.float32)
+    m = oracle.rbq1_mean(X)
+    codes, _, _, _ = oracle.rbq1_encode(X, m)
+    seg = oracle.rbq1_seg_encode(X, m)
+    prep = oracle.rbq1_seg_centroid(C, m)
+    D = oracle.rbq1_seg_partials(codes, seg, d, prep)
+    g = oracle.rbq1_seg_factors(d)
+    assert 0 < g[0] < g[1] < 1
+    prev = r.integers(0, k, n).astype(np.int32)
+    a, est = oracle.rbq1_seg_assign(codes, seg, d, prep, prev=prev)
+    pruned = 0
+    for p in range(n):
+        beta = D[p, prev[p], 2]
+        keep = (D[p, :, 0] <= np.float32(beta * g[0])) & (D[p, :, 1] <= np.float32(beta * g[1]))
+        keep[prev[p]] = True
+        pruned += int((~keep).sum())
+        cand = np.nonzero(keep)[0]
+        want = cand[np.argmin(D[p, cand, 2])]  # np.argmin takes the first (lowest index) on ties
+        assert a[p] == want and est[p] == D[p, want, 2]
+    assert pruned > 0
+    # with no pruning (g = +inf) the result is the argmin of D3 over all centroids
+    a_all, _ = oracle.rbq1_seg_assign(codes, seg, d, prep, prev=prev, g=np.full(2, np.inf, np.float32))
+    np.testing.assert_array_equal(a_all, np.argmin(D[:, :, 2], axis=1))
