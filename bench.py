@@ -635,6 +635,9 @@ def run_case(args):
         pts = skm.rbq1_points(skm.skm_quantize(skm.REPR_RBQ1, X), d)
         if args.case == "assign_rbq1":
             pts = pts.with_screen()
+    elif args.case == "assign_rbq1_skm":  # SuperKMeans checkpoints on RabitQ codes (CUDA cores)
+        q = skm.skm_quantize(skm.REPR_RBQ1, X)
+        pts = skm.rbq1_points(q, d).with_segments(skm.skm_rbq1_segments(X, q["m"])).with_flags(skm.FLAG_PRUNE)
     elif args.case in ("assign_lvq4", "update_lvq4"):
         pts = skm.lvq4_points(skm.skm_quantize(skm.REPR_LVQ4, X), d)
         if args.case == "assign_lvq4":
@@ -661,7 +664,17 @@ def run_case(args):
     wsU = skm.workspace(skm.OP_UPDATE, pts, k)
     a = torch.empty(n, dtype=torch.int32, device="cuda")
     cnt = torch.zeros(k, dtype=torch.int64, device="cuda")
-    skm.skm_assign(pts, C, k, want_dist=False, ws=wsA, out=a)
+    prev = None
+    if args.case == "assign_rbq1_skm":  # the bound from a previous assignment, as in a later Lloyd iteration
+        Cr, _, _, _, _ = skm.skm_fit(pts.with_flags(0), k, 0, init_idx=synth.forgy_indices(n, k, seed=0).cuda(),
+                                     want_objective=False, want_dist=False)
+        C = Cr
+        prev, _ = skm.skm_assign(pts.with_flags(0), C, k, want_dist=False)
+        tp = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        tp[0].record()
+        skm.skm_assign(pts.with_flags(0), C, k, want_dist=False)
+        tp[1].record()
+    skm.skm_assign(pts, C, k, prev_assign=prev, want_dist=False, ws=wsA, out=a)
     torch.cuda.synchronize()
     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     e0.record()
@@ -669,7 +682,7 @@ def run_case(args):
         if args.case == "assign_rbq1_popcount":
             skm.skm_assign_rbq1_noalloc(pts, C, a)
         elif args.case.startswith("assign"):
-            skm.skm_assign(pts, C, k, want_dist=False, ws=wsA, out=a)
+            skm.skm_assign(pts, C, k, prev_assign=prev, want_dist=False, ws=wsA, out=a)
         else:
             skm.skm_update(pts, a, C.clone(), counts=cnt, ws=wsU)
     e1.record()
@@ -679,6 +692,14 @@ def run_case(args):
     if args.case == "assign_f32":  # how often the screen alone decides a row
         _, _, _, _, stats = skm.skm_fit(pts, k, 0, C_init=C, want_objective=False, want_dist=False)
         out["screen_stats"] = stats
+    if args.case == "assign_rbq1_skm":  # survivors per checkpoint, against the dense tensor-core call
+        torch.cuda.synchronize()
+        out["dense_tensor_ms"] = tp[0].elapsed_time(tp[1])
+        _, _, _, _, stats = skm.skm_fit(pts, k, 1, C_init=C, want_objective=False, want_dist=False)
+        pairs = 2.0 * n * k
+        out["after_checkpoint_1"] = stats["prune_first_block"] / pairs
+        out["after_checkpoint_2"] = stats["prune_complete"] / pairs
+        out["same_assignment_as_dense_fraction"] = float((a == prev).float().mean())
     print(json.dumps(out))
 
 
@@ -949,7 +970,8 @@ def main():
     ap.add_argument("--no-extra", action="store_true", help="skip the 1M x 768 and 10M x 1024 1-bit iterations")
     ap.add_argument("--eager", action="store_true", help="time eager steps instead of CUDA-graph replays")
     ap.add_argument("--case", default=None,
-                    help="single-operation run for profiling: assign_f32|assign_bf16|assign_rbq1|assign_sq8|assign_lvq4|"
+                    help="single-operation run for profiling: assign_f32|assign_bf16|assign_rbq1|assign_rbq1_skm|assign_sq8|"
+                         "assign_lvq4|"
                          "assign_rbq1_popcount|assign_prune|assign_prune_sq8|update_f32|update_rbq1|update_sq8|"
                          "update_lvq4|project|quantize_sq8|quantize_rbq1|quantize_lvq4")
     ap.add_argument("--n", type=int, default=200_000)

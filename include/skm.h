@@ -72,7 +72,20 @@ enum {
      * centroid is dropped as soon as its partial distance exceeds the row's
      * current best) instead of the tensor-core path.  Same result (the fp32
      * nearest centroid; for SQ8 the exact integer code-space nearest, with
-     * integer partial sums). */
+     * integer partial sums).
+     * RBQ1, d <= 1024 (with d2 < d, skm_rbq1_segment_bounds): SuperKMeans'
+     * checkpoints for RabitQ codes (Section 3.1): the estimate of Eq.
+     * rabitq_l2 is split over the segments [0, d1), [d1, d2), [d2, d), each
+     * with its own factors (x->seg_*, skm_rbq1_segments) and the centroid's
+     * SQ4 code sums and ||rho_t||^2 per segment, evaluated per segment in the
+     * fp32 order of skm_assign's RBQ1 estimate with fl(1/sqrt(d_t)); partial
+     * estimates D1, D2 and D3 = D2 + est_2 (fp32 sums).  With beta = D3 of
+     * the row's previous centroid (prev_assign; outside [0, k) or NULL:
+     * centroid 0), a centroid other than that one is dropped at checkpoint t
+     * when D_t > fl32(beta g_t), g_t = fl32((e_t / d) (1 + 2.1 / sqrt(e_t))^2)
+     * (ADSampling's scaled test, e_1 = d1, e_2 = d2); the result is the
+     * remaining centroid with the smallest D3, ties to the lowest index, and
+     * dist receives that D3.  AND + popcount on CUDA cores. */
     SKM_FLAG_PRUNE = 1,
     /* RBQ1 only: symmetric 1-bit assignment -- every centroid is binarized
      * like a point (rho = c - m, bit = rho_i > 0) instead of SQ4-coded, and
@@ -108,6 +121,11 @@ typedef struct skm_data {
     /* LVQ4 only (output of skm_quantize): per point (s, b, N, A) of
      * Eq. final:lvq, float32 [n][4], 16-byte aligned                        */
     const float *lvq;
+    /* RBQ1 with SKM_FLAG_PRUNE only (output of skm_rbq1_segments): per point
+     * and dimension segment t = 0, 1, 2: ||r_t||^2, F_t, set bits, [n][3]   */
+    const float *seg_nx2;
+    const float *seg_F;
+    const int32_t *seg_popx;
 } skm_data;
 
 /* Optional per-call statistics (host struct, filled after the call's work
@@ -314,6 +332,20 @@ int skm_column_absmax(const float *X, int64_t n, int d, float *amax_host, void *
 int skm_mean_scale(float amax, int64_t n_total);
 int skm_column_sums_fixed(const float *X, int64_t n, int d, int s, int64_t *sums, void *stream);
 int skm_mean_from_sums(const int64_t *sums, int64_t n_total, int d, int s, float *m, void *stream);
+
+/* SuperKMeans with RabitQ codes (SKM_FLAG_PRUNE on RBQ1): the dimension
+ * segments [0, d1), [d1, d2), [d2, d) with d1 = 32 max(1, floor((d + 128) /
+ * 256)) (12.5% of d in whole 32-dimension words) and d2 = 2 d1; returns
+ * SKM_ERR_UNSUPPORTED when d2 >= d.  Host helper, no GPU use. */
+int skm_rbq1_segment_bounds(int d, int *d1, int *d2);
+
+/* Per point and segment t (r = x - m, the RabitQ mean): nx2s[n][3] =
+ * ||r_t||^2, Fs[n][3] = sqrt(d_t) ||r_t||^2 / ||r_t||_1 (0 when r_t = 0), both
+ * fp64 and rounded once, popxs[n][3] = the set bits of the segment's code
+ * (device outputs; X float32 [n][d], m float32 [d] as given to
+ * skm_quantize).  d <= 1024 with d2 < d.  Asynchronous. */
+int skm_rbq1_segments(const float *X, int64_t n, int d, const float *m, float *nx2s, float *Fs, int32_t *popxs,
+                      void *stream);
 
 /* Fixed-point exponent e of the RBQ1 decode-average: e = 24 - ceil(log2 max F)
  * (0 when every F is 0), so round(F 2^e) <= 2^24 (the largest F keeps its

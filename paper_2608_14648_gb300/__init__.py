@@ -43,7 +43,8 @@ EXPORTED_SYMBOLS = [
     "skm_merge_partials", "skm_update_finalize", "skm_fit", "skm_split_empty", "skm_hier_workspace_size",
     "skm_fit_hierarchical", "skm_objective", "skm_sq8_decode", "skm_step_host_workspace_size",
     "skm_lloyd_step_host", "skm_inject_fault", "skm_fault_armed", "skm_forgy_indices", "skm_column_absmax",
-    "skm_mean_scale", "skm_column_sums_fixed", "skm_mean_from_sums",
+    "skm_mean_scale", "skm_column_sums_fixed", "skm_mean_from_sums", "skm_rbq1_segment_bounds",
+    "skm_rbq1_segments",
 ]
 
 
@@ -61,6 +62,7 @@ class Data(ctypes.Structure):
         ("x", ctypes.c_void_p), ("nx2", ctypes.c_void_p), ("F", ctypes.c_void_p),
         ("popx", ctypes.c_void_p), ("m", ctypes.c_void_p), ("rbq1_exp", ctypes.c_int32),
         ("flags", ctypes.c_int32), ("screen", ctypes.c_void_p), ("lvq", ctypes.c_void_p),
+        ("seg_nx2", ctypes.c_void_p), ("seg_F", ctypes.c_void_p), ("seg_popx", ctypes.c_void_p),
     ]
 
 
@@ -143,6 +145,8 @@ def lib():
             "skm_sq8_decode": ([vp, i64, i32, vp, vp, vp, vp], i32),
             "skm_inject_fault": ([i32, i32], i32),
             "skm_column_absmax": ([vp, i64, i32, vp, vp, sz, vp], i32),
+            "skm_rbq1_segment_bounds": ([i32, vp, vp], i32),
+            "skm_rbq1_segments": ([vp, i64, i32, vp, vp, vp, vp, vp], i32),
             "skm_mean_scale": ([ctypes.c_float, i64], i32),
             "skm_column_sums_fixed": ([vp, i64, i32, i32, vp, vp], i32),
             "skm_mean_from_sums": ([vp, i64, i32, i32, vp, vp], i32),
@@ -186,21 +190,28 @@ class Points:
     """Keeps the tensors of one skm_data alive; `.ref` is the ctypes struct."""
 
     def __init__(self, repr_, x, d, nx2=None, F=None, popx=None, m=None, rbq1_exp=0, screen=None, flags=0,
-                 lvq=None):
+                 lvq=None, seg=None):
         assert x.is_contiguous()
         self.repr, self.x, self.d = repr_, x, int(d)
         self.nx2, self.F, self.popx, self.m = nx2, F, popx, m
         self.lvq = lvq
+        self.seg = seg  # RBQ1 segment factors (nx2s, Fs, popxs), skm_rbq1_segments
         self.n = x.shape[0]
         self.rbq1_exp = int(rbq1_exp)
         self.screen = screen
         self.flags = int(flags)
+        sg = seg if seg is not None else (None, None, None)
         self.ref = Data(repr_, self.d, self.n, x.data_ptr(), _ptr(nx2), _ptr(F), _ptr(popx), _ptr(m),
-                        self.rbq1_exp, self.flags, _ptr(screen), _ptr(lvq))
+                        self.rbq1_exp, self.flags, _ptr(screen), _ptr(lvq), _ptr(sg[0]), _ptr(sg[1]), _ptr(sg[2]))
 
     def with_flags(self, flags):
         return Points(self.repr, self.x, self.d, self.nx2, self.F, self.popx, self.m, self.rbq1_exp, self.screen,
-                      flags, self.lvq)
+                      flags, self.lvq, self.seg)
+
+    def with_segments(self, seg):
+        """The same points with RabitQ segment factors attached (SKM_FLAG_PRUNE on RBQ1)."""
+        return Points(self.repr, self.x, self.d, self.nx2, self.F, self.popx, self.m, self.rbq1_exp, self.screen,
+                      self.flags, self.lvq, seg)
 
     def with_screen(self, stream=None):
         """Builds the screening copy once (skm_screen_prep) and attaches it."""
@@ -210,7 +221,7 @@ class Points:
         buf = _ws(nbytes, self.device)
         _check(lib().skm_screen_prep(ctypes.byref(self.ref), _ptr(buf), buf.numel(), _stream(stream)))
         return Points(self.repr, self.x, self.d, self.nx2, self.F, self.popx, self.m, self.rbq1_exp, buf,
-                      self.flags, self.lvq)
+                      self.flags, self.lvq, self.seg)
 
     @property
     def device(self):
@@ -629,3 +640,20 @@ def skm_mean_from_sums(sums, n_total, s, stream=None):
     m = torch.empty(sums.numel(), device=sums.device, dtype=torch.float32)
     _check(lib().skm_mean_from_sums(_ptr(sums), int(n_total), sums.numel(), int(s), _ptr(m), _stream(stream)))
     return m
+
+
+def skm_rbq1_segment_bounds(d):
+    a, b = ctypes.c_int(0), ctypes.c_int(0)
+    _check(lib().skm_rbq1_segment_bounds(int(d), ctypes.byref(a), ctypes.byref(b)))
+    return a.value, b.value
+
+
+def skm_rbq1_segments(X, m, stream=None):
+    """RabitQ segment factors of the points X (device float32 [n, d]) for the
+    mean m: (nx2s float32 [n, 3], Fs float32 [n, 3], popxs int32 [n, 3])."""
+    n, d = X.shape
+    nx2 = torch.empty(n, 3, device=X.device, dtype=torch.float32)
+    F = torch.empty(n, 3, device=X.device, dtype=torch.float32)
+    pc = torch.empty(n, 3, device=X.device, dtype=torch.int32)
+    _check(lib().skm_rbq1_segments(_ptr(X), n, d, _ptr(m), _ptr(nx2), _ptr(F), _ptr(pc), _stream(stream)))
+    return nx2, F, pc

@@ -90,6 +90,16 @@ static int check_data(const skm_data *x, bool need_codes = true) {
     }
     if ((x->flags & SKM_FLAG_SYMMETRIC) && x->repr != SKM_REPR_RBQ1)
         return set_error(SKM_ERR_INVALID_ARG, "SKM_FLAG_SYMMETRIC applies to RBQ1 only");
+    if ((x->flags & SKM_FLAG_PRUNE) && x->repr == SKM_REPR_RBQ1) {
+        int d1, d2;
+        rbq1_seg_bounds(x->d, &d1, &d2);
+        if (x->d > 1024 || d2 >= x->d)
+            return set_error(SKM_ERR_UNSUPPORTED, "RBQ1 pruning needs 2 d1 < d <= 1024 (d = %d)", x->d);
+        if (x->flags & SKM_FLAG_SYMMETRIC)
+            return set_error(SKM_ERR_UNSUPPORTED, "RBQ1 pruning uses the asymmetric estimate");
+        if (need_codes && (!x->seg_nx2 || !x->seg_F || !x->seg_popx))
+            return set_error(SKM_ERR_INVALID_ARG, "RBQ1 pruning needs the segment factors seg_nx2, seg_F, seg_popx");
+    }
     if (x->repr == SKM_REPR_LVQ4) {
         if (x->n > MAX_N_LVQ4)
             return set_error(SKM_ERR_UNSUPPORTED, "LVQ4 supports n <= 2^26 (got %lld)", (long long)x->n);
@@ -111,8 +121,8 @@ static int check_k(const skm_data *x, int k, bool k_le_n = false) {
 
 // ------------------------------------------------------------ workspace plans
 static bool use_prune(const skm_data *x) {
-    return (x->flags & SKM_FLAG_PRUNE) &&
-           (x->repr == SKM_REPR_F32 || x->repr == SKM_REPR_BF16 || x->repr == SKM_REPR_SQ8);
+    return (x->flags & SKM_FLAG_PRUNE) && (x->repr == SKM_REPR_F32 || x->repr == SKM_REPR_BF16 ||
+                                          x->repr == SKM_REPR_SQ8 || x->repr == SKM_REPR_RBQ1);
 }
 
 struct AssignBufs {
@@ -123,6 +133,7 @@ struct AssignBufs {
     uint32_t *yw = nullptr;                 // LVQ4 with d > 1024 (__dp4a path): centroid nibbles
     float4 *linfo = nullptr;
     TcAssignBufs tc;                        // tensor-core paths (F32, BF16, SQ8, RBQ1)
+    Rbq1SegInfo *seginfo = nullptr;         // RBQ1 with SKM_FLAG_PRUNE (planes above)
 };
 
 static void plan_assign(const skm_data *x, int k, Carver &cv, AssignBufs &b) {
@@ -130,6 +141,10 @@ static void plan_assign(const skm_data *x, int k, Carver &cv, AssignBufs &b) {
     const int d = x->d;
     b.prune = cv.take<unsigned long long>(2);
     if (use_prune(x)) {
+        if (x->repr == SKM_REPR_RBQ1) {
+            b.planes = cv.take<uint4>((size_t)k * words_of(d));
+            b.seginfo = cv.take<Rbq1SegInfo>(k);
+        }
         tc_plan(-1, n, d, k, x->x, x->screen, cv, b.tc);  // statistics only
         return;
     }
@@ -245,6 +260,13 @@ static int do_assign(const skm_data *x, const void *C, int k, const int32_t *pre
     const int64_t n = x->n;
     const int d = x->d;
     if (use_prune(x)) {
+        if (x->repr == SKM_REPR_RBQ1) {
+            SKM_CUDA_TRY(launch_rbq1_seg_cprep(static_cast<const float *>(C), k, d, x->m, b.planes, b.seginfo, st));
+            SKM_CUDA_TRY(launch_assign_rbq1_seg(static_cast<const uint32_t *>(x->x), x->seg_nx2, x->seg_F,
+                                                x->seg_popx, n, d, b.planes, b.seginfo, k, prev, assign, dist,
+                                                b.prune, st));
+            return SKM_OK;
+        }
         if (x->repr == SKM_REPR_SQ8)
             SKM_CUDA_TRY(launch_prune_assign_sq8(static_cast<const uint8_t *>(x->x), n, d, static_cast<const uint8_t *>(C),
                                                  k, prev, assign, dist, b.prune, st));
@@ -670,6 +692,23 @@ int skm_mean_from_sums(const int64_t *sums, int64_t n_total, int d, int s, float
         return set_error(SKM_ERR_INVALID_ARG, "bad shape n=%lld d=%d", (long long)n_total, d);
     SKM_CUDA_TRY(launch_mean_fixed_finish(reinterpret_cast<const unsigned long long *>(sums), d, n_total, nullptr, s,
                                           m, S(stream)));
+    return SKM_OK;
+}
+
+int skm_rbq1_segment_bounds(int d, int *d1, int *d2) {
+    if (!d1 || !d2 || d < 1) return set_error(SKM_ERR_INVALID_ARG, "bad arguments");
+    rbq1_seg_bounds(d, d1, d2);
+    if (*d2 >= d || d > 1024) return set_error(SKM_ERR_UNSUPPORTED, "no segments for d = %d (need 2 d1 < d <= 1024)", d);
+    return SKM_OK;
+}
+
+int skm_rbq1_segments(const float *X, int64_t n, int d, const float *m, float *nx2s, float *Fs, int32_t *popxs,
+                      void *stream) {
+    if (!X || !m || !nx2s || !Fs || !popxs) return set_error(SKM_ERR_INVALID_ARG, "NULL pointer");
+    if (n < 1 || n > MAX_N_RBQ1) return set_error(SKM_ERR_INVALID_ARG, "bad n = %lld", (long long)n);
+    int d1, d2;
+    SKM_TRY(skm_rbq1_segment_bounds(d, &d1, &d2));
+    SKM_CUDA_TRY(launch_rbq1_seg_encode(X, n, d, m, nx2s, Fs, popxs, S(stream)));
     return SKM_OK;
 }
 

@@ -132,6 +132,28 @@ struct Rbq1CInfo {
     float ny2;
 };
 
+// SuperKMeans with RabitQ codes: per-centroid terms of the three dimension
+// segments (SQ4 bias and scale times fl(1/sqrt(d_t)), ||rho_t||^2, code sums)
+struct Rbq1SegInfo {
+    float bd[3];
+    float sd[3];
+    float ny2[3];
+    int32_t sumy[3];
+};
+constexpr double SEG_EPS0 = 2.1;  // ADSampling's significance parameter
+// segments [0, d1), [d1, d2), [d2, d): d1 = d/8 in whole 32-dimension words, d2 = 2 d1
+void rbq1_seg_bounds(int d, int *d1, int *d2);
+// checkpoint factors g_t = fl32((e_t / d) (1 + eps0 / sqrt(e_t))^2)
+void rbq1_seg_factors(int d, int d1, int d2, float *g);
+cudaError_t launch_rbq1_seg_encode(const float *X, int64_t n, int d, const float *m, float *nx2s, float *Fs,
+                                   int32_t *popxs, cudaStream_t st);
+cudaError_t launch_rbq1_seg_cprep(const float *C, int k, int d, const float *m, uint4 *planes, Rbq1SegInfo *info,
+                                  cudaStream_t st);
+cudaError_t launch_assign_rbq1_seg(const uint32_t *codes, const float *nx2s, const float *Fs, const int32_t *popxs,
+                                   int64_t n, int d, const uint4 *planes, const Rbq1SegInfo *info, int k,
+                                   const int32_t *prev, int32_t *assign, float *dist, unsigned long long *counters,
+                                   cudaStream_t st);
+
 // ---- kernels (launchers) ------------------------------------------------
 // quantize / encode
 cudaError_t launch_colminmax_partial(const float *X, int64_t n, int d, float *pmin, float *pmax,

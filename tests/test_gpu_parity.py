@@ -1114,3 +1114,60 @@ def test_sharded_rbq1_mean_codes_and_update_match_single(skm, d):
         skm.skm_merge_partials(total, part)
     C_merged = skm.skm_update_finalize(pw, total, counts, C.clone())
     assert torch.equal(counts, cnt_single) and torch.equal(C_merged, C_single)
+
+
+# ---------------------------------- SuperKMeans with RabitQ codes (checkpoints)
+def _skm_rbq1(skm, n, d, seed):
+    X = _points(n, d, seed=seed).to(DEV)
+    q = skm.skm_quantize(skm.REPR_RBQ1, X)
+    seg = skm.skm_rbq1_segments(X, q["m"])
+    pts = skm.rbq1_points(q, d).with_segments(seg).with_flags(skm.FLAG_PRUNE)
+    return X, q, seg, pts
+
+
+@pytest.mark.parametrize("n,d,k", [(3001, 768, 300), (1000, 1024, 129), (777, 200, 40), (500, 128, 7)])
+def test_rbq1_segment_pruning_bitexact(skm, n, d, k):
+    """Segment factors against the oracle's definitions; the checkpoint-pruned
+    assignment and its D3 equal the oracle's bit for bit (the GPU's factors
+    handed over) for several seeds of the bound."""
+    X, q, seg, pts = _skm_rbq1(skm, n, d, seed=n + d)
+    h = _rbq1_host(q)
+    nx2o, Fo, pco = oracle.rbq1_seg_encode(X.cpu().numpy(), h["m"])
+    segh = tuple(v.cpu().numpy() for v in seg)
+    np.testing.assert_allclose(segh[0], nx2o, rtol=1e-6, atol=1e-12)
+    np.testing.assert_allclose(segh[1], Fo, rtol=1e-6, atol=1e-12)
+    np.testing.assert_array_equal(segh[2], pco)
+    C = X[torch.from_numpy(synth.forgy_indices(n, k, seed=3).numpy()).to(DEV)].clone()
+    C += 0.05 * torch.randn(C.shape, generator=torch.Generator().manual_seed(4)).to(DEV)
+    prep = oracle.rbq1_seg_centroid(C.cpu().numpy(), h["m"])
+    a_plain, _ = skm.skm_assign(skm.rbq1_points(q, d), C)
+    g = torch.Generator().manual_seed(5)
+    for prev in (None, a_plain, torch.randint(0, k, (n,), generator=g, dtype=torch.int32).to(DEV)):
+        a, est = skm.skm_assign(pts, C, prev_assign=prev)
+        ao, esto = oracle.rbq1_seg_assign(h["codes"], segh, d, prep,
+                                          prev=None if prev is None else prev.cpu().numpy())
+        np.testing.assert_array_equal(a.cpu().numpy(), ao)
+        np.testing.assert_array_equal(est.cpu().numpy(), esto)
+
+
+def test_fit_rbq1_segment_pruning_trajectory_bitexact(skm):
+    """skm_fit with the checkpoints (each iteration's bound from the previous
+    assignment) against the oracle's loop of pruned assignments and fused
+    decode-average updates: bit-exact, with pruning statistics reported."""
+    n, d, k, iters = 4000, 256, 60, 4
+    X, q, seg, pts = _skm_rbq1(skm, n, d, seed=77)
+    idx = synth.forgy_indices(n, k, seed=7)
+    C, a, _, _, st = skm.skm_fit(pts, k, iters, init_idx=idx.to(DEV))
+    h = _rbq1_host(q)
+    segh = tuple(v.cpu().numpy() for v in seg)
+    e = pts.rbq1_exp
+    Co = oracle.rbq1_decode_points(h["codes"], h["F"], d, h["m"], e, idx.numpy())
+    prev = None
+    for _ in range(iters):
+        ao, _ = oracle.rbq1_seg_assign(h["codes"], segh, d, oracle.rbq1_seg_centroid(Co, h["m"]), prev=prev)
+        Co, _ = oracle.rbq1_update(h["codes"], h["F"], d, h["m"], e, ao, Co)
+        prev = ao
+    ao, _ = oracle.rbq1_seg_assign(h["codes"], segh, d, oracle.rbq1_seg_centroid(Co, h["m"]), prev=prev)
+    np.testing.assert_array_equal(a.cpu().numpy(), ao)
+    np.testing.assert_array_equal(C.cpu().numpy(), Co)
+    assert 0 < st["prune_complete"] < st["prune_first_block"] < (iters + 1) * n * k
