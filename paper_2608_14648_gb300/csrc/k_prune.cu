@@ -286,6 +286,181 @@ __global__ void __launch_bounds__(PR_WARPS * 32) prune_assign_sq8_kernel(
     }
 }
 
+// ------------------------------------------------------------ tiled kernels
+// A CTA takes TP_PTS points (TP_PTS / 8 per warp) and walks the centroids in
+// chunks of TP_KC staged in shared memory (rows padded so that lanes reading
+// different centroids at the same offset hit different banks), so a chunk
+// is read from L2 once per TP_PTS points instead of once per point.  Per
+// point and chunk, lane l takes the first block of centroids l and l + 32;
+// the survivors are gathered across the warp (ballots, __fns) into dense
+// passes that carry them block by block in lockstep (x's block in registers,
+// read once per pass), leaving as soon as no lane survives.  Each pair's
+// partial sums are the same fp32 (or integer) values as in the kernels above,
+// so the result is the same exact argmin.
+constexpr int TP_PTS = 64;
+constexpr int TP_KC = 64;
+constexpr int TP_WARPS = 8;
+constexpr int TP_MAX_D_F32 = 256;
+
+// sum over the 32 dims of a block: x (registers) against c (shared memory),
+// increasing index order (the order of block_partial)
+__device__ __forceinline__ float block32(const float (&xb)[32], const float *c) {
+    float s = 0.0f;
+#pragma unroll
+    for (int q = 0; q < 8; ++q) {
+        const float4 cv = *reinterpret_cast<const float4 *>(c + 4 * q);
+        float t = __fsub_rn(xb[4 * q], cv.x);
+        s = __fmaf_rn(t, t, s);
+        t = __fsub_rn(xb[4 * q + 1], cv.y);
+        s = __fmaf_rn(t, t, s);
+        t = __fsub_rn(xb[4 * q + 2], cv.z);
+        s = __fmaf_rn(t, t, s);
+        t = __fsub_rn(xb[4 * q + 3], cv.w);
+        s = __fmaf_rn(t, t, s);
+    }
+    return s;
+}
+
+// the i-th survivor of slot masks (M0, M1): slot and owner lane
+__device__ __forceinline__ void survivor(unsigned M0, unsigned M1, int i, int &slot, int &owner) {
+    const int n0 = __popc(M0);
+    slot = i < n0 ? 0 : 1;
+    const unsigned ms = slot == 0 ? M0 : M1;
+    const int rank = slot == 0 ? i : i - n0;
+    owner = (i < n0 + __popc(M1)) ? (int)__fns(ms, 0, rank + 1) : 0;
+}
+
+template <typename TX>
+__global__ void __launch_bounds__(TP_WARPS * 32) prune_tiled_kernel(
+    const TX *__restrict__ X, int64_t n, int d, const float *__restrict__ C, int k,
+    const int32_t *__restrict__ prev, int32_t *__restrict__ assign, float *__restrict__ dist,
+    unsigned long long *__restrict__ counters) {
+    extern __shared__ __align__(16) float tp_smem[];
+    const int dp = ((d + 31) & ~31) + 4;  // padded centroid row (floats): a 16-byte multiple, banks shift by 4
+    const int dx = (d + 31) & ~31;
+    float *cs = tp_smem;                       // [TP_KC][dp]
+    float *xs = cs + (size_t)TP_KC * dp;       // [TP_PTS][dx], zero-padded
+    float *s_beta = xs + (size_t)TP_PTS * dx;  // [TP_PTS]
+    int *s_best = reinterpret_cast<int *>(s_beta + TP_PTS);
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int nb = (d + 31) >> 5;
+    const float slack = 1.0f + 2.0f * (float)(d + 1) * 0x1p-24f;
+    const int64_t p0 = (int64_t)blockIdx.x * TP_PTS;
+    const int np = (int)min((int64_t)TP_PTS, n - p0);
+    unsigned long long first_alive = 0, complete = 0;
+    for (int e = threadIdx.x; e < TP_PTS * dx; e += blockDim.x) {
+        const int q = e / dx, i = e - q * dx;
+        xs[e] = (q < np && i < d) ? ldx<TX>(X + (p0 + q) * d + i) : 0.0f;
+    }
+    __syncthreads();
+    // each point's bound: its full distance to the seed centroid (block sums in order)
+    for (int q = warp; q < np; q += TP_WARPS) {
+        int best = prev ? prev[p0 + q] : 0;
+        if (best < 0 || best >= k) best = 0;
+        if (lane == 0) {
+            float beta = 0.0f;
+            for (int b = 0; b < nb; ++b) beta += block_partial(xs + q * dx, C + (int64_t)best * d, d, b);
+            s_beta[q] = beta;
+            s_best[q] = best;
+        }
+    }
+    for (int c0 = 0; c0 < k; c0 += TP_KC) {
+        const int kc = min(TP_KC, k - c0);
+        __syncthreads();
+        for (int e = threadIdx.x; e < TP_KC * dx; e += blockDim.x) {
+            const int c = e / dx, i = e - c * dx;
+            cs[c * dp + i] = (c < kc && i < d) ? C[(int64_t)(c0 + c) * d + i] : 0.0f;
+        }
+        __syncthreads();
+        for (int q = warp; q < np; q += TP_WARPS) {
+            const float *xq = xs + q * dx;
+            float beta = s_beta[q];
+            int best = s_best[q];
+            float lim = beta * slack;
+            float xb[32];
+#pragma unroll
+            for (int u = 0; u < 8; ++u) {
+                const float4 v = *reinterpret_cast<const float4 *>(xq + 4 * u);  // broadcast
+                xb[4 * u] = v.x;
+                xb[4 * u + 1] = v.y;
+                xb[4 * u + 2] = v.z;
+                xb[4 * u + 3] = v.w;
+            }
+            float pa[2];
+            unsigned M[2];
+#pragma unroll
+            for (int s2 = 0; s2 < 2; ++s2) {
+                const int c = 32 * s2 + lane;
+                // a partial block past d sums zeros (both sides padded), as block_partial
+                pa[s2] = c < kc ? block32(xb, cs + c * dp) : INFINITY;
+                M[s2] = __ballot_sync(0xffffffffu, c < kc && pa[s2] <= lim);
+            }
+            const int total = __popc(M[0]) + __popc(M[1]);
+            first_alive += lane == 0 ? (unsigned long long)total : 0ull;
+            for (int base = 0; base < total; base += 32) {
+                const int i = base + lane;
+                int slot, owner;
+                survivor(M[0], M[1], i, slot, owner);
+                const float v0 = __shfl_sync(0xffffffffu, pa[0], owner);
+                const float v1 = __shfl_sync(0xffffffffu, pa[1], owner);
+                const bool mine = i < total;
+                const int c = 32 * slot + owner;
+                float p = slot == 0 ? v0 : v1;
+                bool alive = mine;
+                for (int b = 1; b < nb; ++b) {
+                    if (!__any_sync(0xffffffffu, alive)) break;
+#pragma unroll
+                    for (int u = 0; u < 8; ++u) {
+                        const float4 v = *reinterpret_cast<const float4 *>(xq + 32 * b + 4 * u);
+                        xb[4 * u] = v.x;
+                        xb[4 * u + 1] = v.y;
+                        xb[4 * u + 2] = v.z;
+                        xb[4 * u + 3] = v.w;
+                    }
+                    if (alive) {
+                        p += block32(xb, cs + c * dp + 32 * b);
+                        alive = p <= lim;
+                    }
+                }
+                complete += alive ? 1ull : 0ull;
+                float bp = alive ? p : INFINITY;
+                int bj = alive ? c0 + c : 0x7fffffff;
+#pragma unroll
+                for (int o = 16; o > 0; o >>= 1) {
+                    const float op = __shfl_xor_sync(0xffffffffu, bp, o);
+                    const int oj = __shfl_xor_sync(0xffffffffu, bj, o);
+                    if (op < bp || (op == bp && oj < bj)) {
+                        bp = op;
+                        bj = oj;
+                    }
+                }
+                if (bp < beta || (bp == beta && bj < best)) {
+                    beta = bp;
+                    best = bj;
+                    lim = beta * slack;
+                }
+            }
+            if (lane == 0) {
+                s_beta[q] = beta;
+                s_best[q] = best;
+            }
+        }
+    }
+    __syncthreads();
+    for (int q = threadIdx.x; q < np; q += blockDim.x) {
+        assign[p0 + q] = s_best[q];
+        if (dist) dist[p0 + q] = s_beta[q];
+    }
+    if (counters) {
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) complete += __shfl_xor_sync(0xffffffffu, complete, o);
+        if (lane == 0) {
+            atomicAdd(&counters[0], first_alive);
+            atomicAdd(&counters[1], complete);
+        }
+    }
+}
+
 }  // namespace
 
 cudaError_t launch_prune_assign_sq8(const uint8_t *X, int64_t n, int d, const uint8_t *C, int k, const int32_t *prev,
@@ -301,6 +476,25 @@ cudaError_t launch_prune_assign(const void *X, int x_is_bf16, int64_t n, int d, 
                                 int k, const int32_t *prev, int32_t *assign, float *dist,
                                 unsigned long long *counters, cudaStream_t st) {
     if (n == 0) return cudaSuccess;
+    if (d <= TP_MAX_D_F32 && (reinterpret_cast<uintptr_t>(C) & 15) == 0) {
+        const int dx = (d + 31) & ~31, dp = dx + 4;
+        const size_t smem = ((size_t)TP_KC * dp + (size_t)TP_PTS * dx + 2 * TP_PTS) * sizeof(float);
+        const int64_t blocks = (n + TP_PTS - 1) / TP_PTS;
+        if (x_is_bf16) {
+            cudaError_t e = cudaFuncSetAttribute(prune_tiled_kernel<uint16_t>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                                 (int)smem);
+            if (e != cudaSuccess) return e;
+            prune_tiled_kernel<uint16_t><<<(unsigned)blocks, TP_WARPS * 32, smem, st>>>(
+                static_cast<const uint16_t *>(X), n, d, C, k, prev, assign, dist, counters);
+        } else {
+            cudaError_t e = cudaFuncSetAttribute(prune_tiled_kernel<float>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                                 (int)smem);
+            if (e != cudaSuccess) return e;
+            prune_tiled_kernel<float><<<(unsigned)blocks, TP_WARPS * 32, smem, st>>>(
+                static_cast<const float *>(X), n, d, C, k, prev, assign, dist, counters);
+        }
+        return launched();
+    }
     int64_t blocks = (n + PR_WARPS - 1) / PR_WARPS;
     if (blocks > 152 * 16) blocks = 152 * 16;
     if (x_is_bf16)
