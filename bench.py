@@ -47,13 +47,27 @@ POPC_PER_CLK_SM = 16
 # DRAM bytes (read + write) per point of the assignment kernels, each from
 # one ncu capture of a smaller case of the same kernel (every point row is
 # read once per launch, so traffic scales with the points): the bf16 screen
-# at 400,000 x 256 with k = 10,000; the fp32 screen and the e4m3 1-bit
-# kernel at 200,000 x 768 with k = 1,000.
+# at 400,000 x 256 with k = 10,000; the fp32 screen and the 1-bit kernel
+# (packed codes, tiles expanded in an L2-resident scratch) at 200,000 x 768
+# with k = 1,000.
 TRAFFIC_PER_POINT = {
     "assign_bf16_screen": (213.449216e6 + 4.711680e6) / 400_000,
     "assign_f32": (314.849280e6 + 5.701888e6) / 200_000,
-    "assign_rbq1": (156.890624e6 + 3.590912e6) / 200_000,
+    "assign_rbq1": (22.462464e6 + 23.388416e6) / 200_000,
 }
+
+
+def prune_roofline(pairs, later_blocks, nb, ms, peaks):
+    """Executed-work roofline of a pruned assignment: every (point, centroid)
+    pair's first 32-dimension block plus the later blocks the bounds did not
+    skip, each 32 fp32 subtractions and 32 fmas on the CUDA cores, against
+    SM_COUNT SMs x 128 fp32 lanes at the maximum SM clock."""
+    blocks = pairs + float(later_blocks)
+    achieved = blocks * 64.0 / (ms / 1e3) / 1e12
+    peak = SM_COUNT * 128 * peaks["sm_max_mhz"] * 1e6 / 1e12
+    return {"bound": "alu", "unit": "T fp32 lane-instructions/s", "executed_blocks": blocks,
+            "executed_fraction_of_dense": blocks / (pairs * nb), "achieved": achieved, "peak": peak,
+            "frac": achieved / peak}
 
 
 def env_rank():
@@ -290,7 +304,7 @@ def run_extra_configs(args, dev, peaks, stream, local_rank):
 
     out = {}
 
-    def timed(name, pts, C, k, n, d, flop_peak, kind):
+    def timed(name, pts, C, k, n, d, flop_peak, kind, copy_pts=None):
         wsA = skm.workspace(skm.OP_ASSIGN, pts, k)
         wsU = skm.workspace(skm.OP_UPDATE, pts, k)
         a = torch.empty(n, dtype=torch.int32, device=dev)
@@ -310,6 +324,13 @@ def run_extra_configs(args, dev, peaks, stream, local_rank):
                      "assign_ms": t_a, "update_ms": t_u, "assign_achieved_tflops": ach, "assign_peak_tflops": flop_peak,
                      "assign_frac": ach / flop_peak, "flop": kind, "steps": steps, "timing": timing, "clocks": clk,
                      "gpu_launches": launches}
+        if copy_pts is not None:  # 1-bit: the points stay packed; the e4m3 copy for comparison
+            wsC = skm.workspace(skm.OP_ASSIGN, copy_pts, k)
+            t_c = _event_ms(lambda: skm.skm_assign(copy_pts, C, k, want_dist=False, ws=wsC, out=a), 3, stream)
+            out[name]["points_in_hbm"] = f"packed 1-bit codes, {4 * ((d + 31) // 32)} B a point"
+            out[name]["assign_ms_from_e4m3_copy"] = t_c
+            out[name]["e4m3_copy_bytes"] = n * (d + 15) // 16 * 16
+            del wsC
         del wsA, wsU
 
     bf16 = peaks["bf16_tflops"]
@@ -318,9 +339,9 @@ def run_extra_configs(args, dev, peaks, stream, local_rank):
     idx = synth.forgy_indices(spec.n, spec.k, seed=0).to(dev)
     timed("emb1m_d768_f32", skm.Points(skm.REPR_F32, X, spec.d).with_screen(), X[idx].clone(), spec.k, spec.n,
           spec.d, bf16, "bf16")
-    pR = skm.rbq1_points(skm.skm_quantize(skm.REPR_RBQ1, X), spec.d).with_screen()
+    pR = skm.rbq1_points(skm.skm_quantize(skm.REPR_RBQ1, X), spec.d)
     CR, _, _, _, _ = skm.skm_fit(pR, spec.k, 0, init_idx=idx, want_objective=False, want_dist=False)
-    timed("emb1m_d768_rbq1", pR, CR, spec.k, spec.n, spec.d, 2 * bf16, "e4m3")
+    timed("emb1m_d768_rbq1", pR, CR, spec.k, spec.n, spec.d, 2 * bf16, "e4m3", copy_pts=pR.with_screen())
     # the AND + popcount 1-bit kernel on the same codes (no allocation entry point)
     a_pop = torch.empty(spec.n, dtype=torch.int32, device=dev)
     skm.skm_assign_rbq1_noalloc(pR, CR, a_pop)
@@ -342,9 +363,9 @@ def run_extra_configs(args, dev, peaks, stream, local_rank):
     del Y
     torch.cuda.empty_cache()
     idx = synth.forgy_indices(spec.n, spec.k, seed=0).to(dev)
-    pR = skm.rbq1_points(q, spec.d).with_screen()
+    pR = skm.rbq1_points(q, spec.d)
     CR, _, _, _, _ = skm.skm_fit(pR, spec.k, 0, init_idx=idx, want_objective=False, want_dist=False)
-    timed("emb10m_d1024_rbq1", pR, CR, spec.k, spec.n, spec.d, 2 * bf16, "e4m3")
+    timed("emb10m_d1024_rbq1", pR, CR, spec.k, spec.n, spec.d, 2 * bf16, "e4m3", copy_pts=pR.with_screen())
     del pR, CR, q
     torch.cuda.empty_cache()
     return out
@@ -425,16 +446,17 @@ def run_ours(args):
         skm.skm_assign(pp, C_step, K, prev_assign=prev, want_dist=False, ws=wsP, out=ap)
         t_prune = _event_ms(lambda: skm.skm_assign(pp, C_step, K, prev_assign=prev, want_dist=False, ws=wsP,
                                                    out=ap), 2, stream)
-        _, _, _, _, st = skm.skm_fit(pp, K, 0, C_init=C_step, want_objective=False, want_dist=False)
+        st = skm.skm_assign_prune_stats(wsP, stream)  # counters of the last timed call
         same = bool(torch.equal(ap, a[:ns]))
         pairs = float(ns) * K
         dense_ms = t_assign * ns / N
         kernels["assign_bf16_prune"] = {
-            "ms": t_prune, "rows": ns, "in_step": False, "bound": "fp32 CUDA cores",
+            "ms": t_prune, "rows": ns, "in_step": False,
             "first_block_survivors": st["prune_first_block"] / pairs, "complete_survivors": st["prune_complete"] / pairs,
             "dense_screen_ms_same_rows": dense_ms, "speedup_vs_dense": dense_ms / t_prune,
             "same_assignment_as_dense": same,
-            "note": "exact 32-dimension prefix-block pruning, bound seeded with the previous assignment"}
+            "note": "exact 32-dimension prefix-block pruning, bound seeded with the previous assignment",
+            **prune_roofline(pairs, st["prune_blocks"], D_PCA // 32, t_prune, peaks)}
         del pp, ap, prev, wsP
     for kd in kernels.values():
         if "achieved" in kd:
@@ -633,7 +655,7 @@ def run_case(args):
         pts = skm.Points(skm.REPR_F32, X, d).with_screen()
     elif args.case in ("assign_rbq1", "update_rbq1", "assign_rbq1_popcount"):
         pts = skm.rbq1_points(skm.skm_quantize(skm.REPR_RBQ1, X), d)
-        if args.case == "assign_rbq1":
+        if args.case == "assign_rbq1" and args.e4m3_copy:  # the e4m3 screening copy instead of packed codes
             pts = pts.with_screen()
     elif args.case == "assign_rbq1_skm":  # SuperKMeans checkpoints on RabitQ codes (CUDA cores)
         q = skm.skm_quantize(skm.REPR_RBQ1, X)
@@ -689,6 +711,12 @@ def run_case(args):
     torch.cuda.synchronize()
     out = {"case": args.case, "n": n, "d": d, "k": k, "reps": args.reps,
            "ms_per_call": e0.elapsed_time(e1) / args.reps}
+    if args.case in ("assign_prune", "assign_prune_sq8"):  # the work the bounds left (last timed call)
+        st = skm.skm_assign_prune_stats(wsA)
+        pairs = float(n) * k
+        out["first_block_survivors"] = st["prune_first_block"] / pairs
+        out["complete_survivors"] = st["prune_complete"] / pairs
+        out["later_blocks_per_pair"] = st["prune_blocks"] / pairs
     if args.case == "assign_f32":  # how often the screen alone decides a row
         _, _, _, _, stats = skm.skm_fit(pts, k, 0, C_init=C, want_objective=False, want_dist=False)
         out["screen_stats"] = stats
@@ -975,6 +1003,8 @@ def main():
                          "assign_rbq1_popcount|assign_prune|assign_prune_sq8|update_f32|update_rbq1|update_sq8|"
                          "update_lvq4|project|quantize_sq8|quantize_rbq1|quantize_lvq4")
     ap.add_argument("--n", type=int, default=200_000)
+    ap.add_argument("--e4m3-copy", action="store_true",
+                    help="--case assign_rbq1: read the points from their e4m3 copy instead of packed")
     ap.add_argument("--d", type=int, default=768)
     ap.add_argument("--k", type=int, default=1000)
     ap.add_argument("--reps", type=int, default=3)

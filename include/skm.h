@@ -144,7 +144,11 @@ typedef struct skm_stats {
                                  entries, or NULL; skm_fit writes the number of
                                  empty clusters after each update (before any
                                  split) of its first 4096 iterations           */
-    int64_t reserved;
+    int64_t prune_blocks;     /* SKM_FLAG_PRUNE on F32/BF16/SQ8: 32-dimension
+                                 block partial sums evaluated after the first
+                                 block (the executed work beyond the n k first
+                                 blocks); 0 for RBQ1, whose checkpoints are
+                                 counted by the two fields above               */
 } skm_stats;
 
 const char *skm_last_error(void);
@@ -369,7 +373,15 @@ int skm_lvq4_exponent(const float *lvq, int64_t n, int *e_host, void *ws, size_t
  * -> the codes as e4m3 bytes.  skm_screen_bytes returns its size (0 when the
  * representation needs none: SQ8, RBQ1 or LVQ4 with d > 1024);
  * skm_screen_prep fills `screen` (device, 256-byte aligned,
- * caller-owned) from x->x.  Asynchronous. */
+ * caller-owned) from x->x.  Asynchronous.
+ * RBQ1 without a copy (x->screen NULL): when a code row is a multiple of 16
+ * bytes (ceil(d/32) a multiple of 4) at a 16-byte aligned address, the
+ * assignment reads the codes packed (each CTA expands its point tiles into a
+ * slot of the workspace, at most 160 x 4 x 128 x round16(d) bytes), so the
+ * points occupy ceil(d/32) words in HBM instead of round16(d) bytes; the copy
+ * saves that per-tile expansion (measured on GB300: 1M x 768, k = 1000: 0.61
+ * ms packed, 0.53 ms from the copy).  Otherwise skm_assign builds the copy in
+ * its workspace on every call. */
 size_t skm_screen_bytes(const skm_data *x);
 int skm_screen_prep(const skm_data *x, void *screen, size_t screen_bytes, void *stream);
 
@@ -416,6 +428,17 @@ int skm_screen_prep(const skm_data *x, void *screen, size_t screen_bytes, void *
  * ------------------------------------------------------------------------ */
 int skm_assign(const skm_data *x, const void *C, int k, const int32_t *prev_assign,
                int32_t *assign, float *dist, void *ws, size_t ws_bytes, void *stream);
+
+/* Pruning counters of the last skm_assign call with SKM_FLAG_PRUNE that ran
+ * on workspace `ws` (Section 3.1 "SuperKMeans": the work the bounds skipped).
+ * skm_assign zeroes them at the start of such a call.  Fills
+ * prune_first_block, prune_complete and prune_blocks of *out (the other
+ * fields are zero); for RBQ1 the first two count the pairs alive after the
+ * 12.5% and 25% checkpoints.  Synchronises `stream` (the caller's device
+ * pointer `ws`, at least the size skm_workspace_size returned for that call).
+ * Errors: SKM_ERR_INVALID_ARG (NULL ws or out, ws_bytes too small for the
+ * counters), SKM_ERR_CUDA. */
+int skm_assign_prune_stats(const void *ws, size_t ws_bytes, skm_stats *out, void *stream);
 
 /* RBQ1 assignment that allocates nothing.  The paper has no counterpart:
  * this entry point exists for callers that cannot allocate device memory

@@ -20,6 +20,7 @@ __all__ = [
     "skm_quantize", "skm_rbq1_exponent", "skm_lvq4_exponent", "skm_assign", "skm_update", "skm_merge_partials",
     "skm_update_finalize", "skm_fit", "skm_split_empty", "skm_objective", "skm_sq8_decode", "EXPORTED_SYMBOLS",
     "EMPTY_KEEP", "EMPTY_SPLIT",
+    "skm_assign_prune_stats",
 ]
 
 REPR_F32, REPR_SQ8, REPR_RBQ1, REPR_BF16, REPR_LVQ4 = 0, 1, 2, 3, 4
@@ -37,7 +38,8 @@ EXPORTED_SYMBOLS = [
     "skm_last_error", "skm_version", "skm_kernel_launches", "skm_workspace_size", "skm_screen_bytes",
     "skm_screen_prep", "skm_project", "skm_project_hadamard", "skm_unproject", "skm_copy_from_host",
     "skm_make_rotation",
-    "skm_pca_fit", "skm_quantize", "skm_rbq1_exponent", "skm_lvq4_exponent", "skm_assign", "skm_assign_rbq1_noalloc",
+    "skm_pca_fit", "skm_quantize", "skm_rbq1_exponent", "skm_lvq4_exponent", "skm_assign",
+    "skm_assign_prune_stats", "skm_assign_rbq1_noalloc",
     "skm_assign_segmented",
     "skm_update",
     "skm_merge_partials", "skm_update_finalize", "skm_fit", "skm_split_empty", "skm_hier_workspace_size",
@@ -78,7 +80,7 @@ class Stats(ctypes.Structure):
     _fields_ = [("rescored_rows", ctypes.c_int64), ("fallback_rows", ctypes.c_int64),
                 ("empty_clusters", ctypes.c_int64), ("prune_first_block", ctypes.c_int64),
                 ("prune_complete", ctypes.c_int64), ("cluster_size_std", ctypes.c_double),
-                ("empty_per_iter", ctypes.c_void_p), ("reserved", ctypes.c_int64)]
+                ("empty_per_iter", ctypes.c_void_p), ("prune_blocks", ctypes.c_int64)]
 
 
 class HierConfig(ctypes.Structure):
@@ -132,6 +134,7 @@ def lib():
             "skm_rbq1_exponent": ([vp, i64, vp, vp, sz, vp], i32),
             "skm_lvq4_exponent": ([vp, i64, vp, vp, sz, vp], i32),
             "skm_assign": ([vp, vp, i32, vp, vp, vp, vp, sz, vp], i32),
+            "skm_assign_prune_stats": ([vp, sz, vp, vp], i32),
             "skm_assign_rbq1_noalloc": ([vp, vp, i32, vp, vp, vp], i32),
             "skm_assign_segmented": ([vp, vp, i32, vp, vp, i32, vp, vp, vp, sz, vp], i32),
             "skm_update": ([vp, vp, i32, vp, vp, vp, vp, sz, vp], i32),
@@ -415,6 +418,16 @@ def skm_assign(pts: Points, C, k=None, prev_assign=None, want_dist=True, ws=None
     return assign, dist
 
 
+def skm_assign_prune_stats(ws, stream=None):
+    """Pruning counters of the last pruned skm_assign on workspace `ws`
+    (synchronises the stream): first-block / complete survivors and the
+    block partial sums evaluated after the first block."""
+    st = Stats()
+    _check(lib().skm_assign_prune_stats(_ptr(ws), ws.numel(), ctypes.byref(st), _stream(stream)))
+    return {"prune_first_block": st.prune_first_block, "prune_complete": st.prune_complete,
+            "prune_blocks": st.prune_blocks}
+
+
 def skm_assign_rbq1_noalloc(pts: Points, C, out, dist_out=None, stream=None):
     """RBQ1 assignment that allocates nothing in the library (fixed device
     scratch); `out` (int32[n]) and `dist_out` (float[n] or None) are caller
@@ -499,7 +512,8 @@ def skm_fit(pts: Points, k, iters, C_init=None, init_idx=None, want_objective=Tr
                          _ptr(assign), _ptr(dist), obj, ctypes.byref(st), _ptr(ws), ws.numel(), _stream(stream)))
     stats = {"rescored_rows": st.rescored_rows, "fallback_rows": st.fallback_rows,
              "empty_clusters": st.empty_clusters, "prune_first_block": st.prune_first_block,
-             "prune_complete": st.prune_complete, "cluster_size_std": st.cluster_size_std,
+             "prune_complete": st.prune_complete, "prune_blocks": st.prune_blocks,
+             "cluster_size_std": st.cluster_size_std,
              "empty_per_iter": list(empties)[:min(iters, 4096)]}
     return C, assign, dist, (list(obj) if obj is not None else None), stats
 

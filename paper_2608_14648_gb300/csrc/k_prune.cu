@@ -78,7 +78,7 @@ __global__ void __launch_bounds__(PR_WARPS * 32) prune_assign_kernel(
     // d * 2^-24; keep anything within twice that of beta
     const float slack = 1.0f + 2.0f * (float)(d + 1) * 0x1p-24f;
     const int64_t nw = (int64_t)gridDim.x * PR_WARPS;
-    unsigned long long first_alive = 0, complete = 0;
+    unsigned long long first_alive = 0, complete = 0, later = 0;
     for (int64_t row = (int64_t)blockIdx.x * PR_WARPS + warp; row < n; row += nw) {
         __syncwarp();
         for (int i = lane; i < d; i += 32) sx[i] = ldx<TX>(X + row * d + i);
@@ -107,6 +107,7 @@ __global__ void __launch_bounds__(PR_WARPS * 32) prune_assign_kernel(
             int src = 0;
             for (int b = 1; b < nb && cnt > 0; ++b) {
                 __syncwarp();
+                later += cnt;
                 int ncnt = 0;
                 for (int t0 = 0; t0 < cnt; t0 += 32) {
                     const int t = t0 + lane;
@@ -160,6 +161,7 @@ __global__ void __launch_bounds__(PR_WARPS * 32) prune_assign_kernel(
     if (counters && lane == 0) {
         atomicAdd(&counters[0], first_alive);
         atomicAdd(&counters[1], complete);
+        atomicAdd(&counters[2], later);
     }
 }
 
@@ -204,7 +206,7 @@ __global__ void __launch_bounds__(PR_WARPS * 32) prune_assign_sq8_kernel(
     const int nb = (d + 31) >> 5;
     const bool words = (d % 4) == 0 && (reinterpret_cast<uintptr_t>(C) & 3) == 0;
     const int64_t nw = (int64_t)gridDim.x * PR_WARPS;
-    unsigned long long first_alive = 0, complete = 0;
+    unsigned long long first_alive = 0, complete = 0, later = 0;
     for (int64_t row = (int64_t)blockIdx.x * PR_WARPS + warp; row < n; row += nw) {
         __syncwarp();
         for (int i = lane; i < d; i += 32) sx[i] = __ldg(X + row * d + i);
@@ -232,6 +234,7 @@ __global__ void __launch_bounds__(PR_WARPS * 32) prune_assign_sq8_kernel(
             int src = 0;
             for (int b = 1; b < nb && cnt > 0; ++b) {
                 __syncwarp();
+                later += cnt;
                 int ncnt = 0;
                 for (int t0 = 0; t0 < cnt; t0 += 32) {
                     const int t = t0 + lane;
@@ -283,6 +286,7 @@ __global__ void __launch_bounds__(PR_WARPS * 32) prune_assign_sq8_kernel(
     if (counters && lane == 0) {
         atomicAdd(&counters[0], first_alive);
         atomicAdd(&counters[1], complete);
+        atomicAdd(&counters[2], later);
     }
 }
 
@@ -347,7 +351,7 @@ __global__ void __launch_bounds__(TP_WARPS * 32) prune_tiled_kernel(
     const float slack = 1.0f + 2.0f * (float)(d + 1) * 0x1p-24f;
     const int64_t p0 = (int64_t)blockIdx.x * TP_PTS;
     const int np = (int)min((int64_t)TP_PTS, n - p0);
-    unsigned long long first_alive = 0, complete = 0;
+    unsigned long long first_alive = 0, complete = 0, later = 0;
     for (int e = threadIdx.x; e < TP_PTS * dx; e += blockDim.x) {
         const int q = e / dx, i = e - q * dx;
         xs[e] = (q < np && i < d) ? ldx<TX>(X + (p0 + q) * d + i) : 0.0f;
@@ -420,6 +424,7 @@ __global__ void __launch_bounds__(TP_WARPS * 32) prune_tiled_kernel(
                     if (alive) {
                         p += block32(xb, cs + c * dp + 32 * b);
                         alive = p <= lim;
+                        ++later;
                     }
                 }
                 complete += alive ? 1ull : 0ull;
@@ -453,10 +458,14 @@ __global__ void __launch_bounds__(TP_WARPS * 32) prune_tiled_kernel(
     }
     if (counters) {
 #pragma unroll
-        for (int o = 16; o > 0; o >>= 1) complete += __shfl_xor_sync(0xffffffffu, complete, o);
+        for (int o = 16; o > 0; o >>= 1) {
+            complete += __shfl_xor_sync(0xffffffffu, complete, o);
+            later += __shfl_xor_sync(0xffffffffu, later, o);
+        }
         if (lane == 0) {
             atomicAdd(&counters[0], first_alive);
             atomicAdd(&counters[1], complete);
+            atomicAdd(&counters[2], later);
         }
     }
 }

@@ -52,6 +52,15 @@ constexpr int BK = 64;   // bf16 elements per 128-byte swizzle row
 constexpr int STAGES = 4;
 constexpr int A_STAGE = BM * BK * 2;  // 16 KiB
 constexpr int B_STAGE = BN * BK * 2;  // 32 KiB
+// 1-bit points kept packed in HBM: CONV_WARPS converter warps expand each of
+// a CTA's point tiles once, a tile ahead of the producer, into that CTA's
+// scratch in global memory (two slots per job stream, 128 rows of round16(d)
+// e4m3 bytes each: at most PK_MAX_CTAS x 2 x 2 x 128 KiB, which L2 keeps),
+// from where the TMA loads the A slices exactly as from an e4m3 copy of all
+// the points.  The conversion is paid once per point tile instead of once
+// per (point tile, centroid tile) job.
+constexpr int CONV_WARPS = 4;
+constexpr int PK_MAX_CTAS = 160;
 constexpr int TCAND = 4;
 constexpr unsigned long long WAIT_LIMIT_NS = 2000000000ull;  // 2 s per barrier wait
 
@@ -93,8 +102,8 @@ constexpr bool f8_mode() { return MODE == MODE_RBQ1 || MODE == MODE_LVQ4; }
 // Epilogue shape: NH warps per TMEM lane quarter (column slices of 256 / NH).
 template <int NH>
 constexpr int epi_threads() { return 128 * NH; }
-template <int NH>
-constexpr int tc_threads() { return 64 + epi_threads<NH>(); }
+template <int NH, bool PK = false>
+constexpr int tc_threads() { return 64 + epi_threads<NH>() + (PK ? 32 * CONV_WARPS : 0); }
 // one row's state for the merge: the screen list, or (best, index)
 template <int MODE>
 constexpr int merge_words() { return MODE == MODE_SCREEN ? 2 * TCAND + 2 : 2; }
@@ -136,6 +145,11 @@ struct TcParams {
     const float4 *lvq;       // LVQ4 per point (s, b, N, A); rinfo / rinfoq hold
                              // the column pairs (b x2, G x2) / (s x2, N x2)
     int d;
+    // RBQ1 read packed: the codes [n][pk_words] and the CTAs' expansion
+    // scratch (slot ((cta NS + stream) 2 + i) of BM x pk_dp bytes)
+    const uint32_t *pk_codes;
+    uint8_t *pk_scratch;
+    int pk_words, pk_dp;
     // Segmented mode (all NULL otherwise): the point rows are sorted by
     // group and row r may only take centroids [seg_base[g], seg_base[g + 1])
     // of its group g = seg_group[r]; point tile rt covers the centroid tiles
@@ -314,6 +328,14 @@ __device__ __forceinline__ float2 fmul2(float2 a, float2 b) {
     return r;
 }
 
+// Bits 0..3 of v -> four e4m3 bytes, bit j -> byte j: +1.0 (0x38) when set,
+// -1.0 (0xB8) when clear.  The product puts bit j of the nibble at bit 8j + 7
+// (the partial products land on distinct bits, so nothing carries).
+__device__ __forceinline__ uint32_t pm1_e4m3(uint32_t v) {
+    const uint32_t t = (v & 15u) * 0x10204080u;
+    return (t & 0x80808080u) ^ 0xB8B8B8B8u;
+}
+
 // min(a, b, c) in one instruction (sm_100 family three-input min)
 __device__ __forceinline__ float fmin3(float a, float b, float c) {
     float r;
@@ -440,8 +462,8 @@ __device__ __forceinline__ void ct_range(const TcParams &p, int64_t rt, int &lo,
     }
 }
 
-template <int MODE, int NH, bool SEG, int NS>
-__global__ void __launch_bounds__(tc_threads<NH>(), 1)
+template <int MODE, int NH, bool SEG, int NS, bool PK>
+__global__ void __launch_bounds__(tc_threads<NH, PK>(), 1)
     tc_assign_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                      const TcParams p) {
     static_assert(NS == 1 || (NS == 2 && NH % 2 == 0), "two job streams: two epilogue groups");
@@ -464,6 +486,12 @@ __global__ void __launch_bounds__(tc_threads<NH>(), 1)
     // the injected wait (nothing arrives on either otherwise)
     const uint32_t drain_bar = bar0 + 8u * (2 * STAGES + 5);
     const uint32_t inject_bar = bar0 + 8u * (2 * STAGES + 6);
+    // PK: scratch slot i of job stream j is written (count: one arrival per
+    // converter warp) / free again (the MMA warp, once the last TMA load
+    // from it has landed)
+    auto sready_bar = [&](int j, int i) { return bar0 + 8u * (2 * STAGES + 7 + 2 * j + i); };
+    auto sfree_bar = [&](int j, int i) { return bar0 + 8u * (2 * STAGES + 11 + 2 * j + i); };
+    static_assert(!PK || MODE == MODE_RBQ1, "packed points: 1-bit codes only");
     // the epilogue's merge buffer starts 256 bytes after tmem_slot (see tc_smem_bytes)
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -482,6 +510,12 @@ __global__ void __launch_bounds__(tc_threads<NH>(), 1)
         }
         mbar_init(drain_bar, 1);
         mbar_init(inject_bar, 1);
+        if (PK)
+            for (int j = 0; j < NS; ++j)
+                for (int i = 0; i < 2; ++i) {
+                    mbar_init(sready_bar(j, i), CONV_WARPS);
+                    mbar_init(sfree_bar(j, i), 1);
+                }
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
         asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmA)) : "memory");
         asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmB)) : "memory");
@@ -553,8 +587,12 @@ __global__ void __launch_bounds__(tc_threads<NH>(), 1)
             if (p.inject_wait_ns && !mbar_wait(inject_bar, 0u, abort_flag, p.inject_wait_ns)) goto producer_done;
             {
             JobStream js[NS];
+            int64_t ptile[NS];  // PK: each stream's current point tile and tiles taken
+            uint32_t pcnt[NS];
             for (int s = 0; s < NS; ++s) {
                 js[s].g = g0 + s * gstep;
+                ptile[s] = -1;
+                pcnt[s] = 0;
                 stream_seek(js[s]);
             }
             for (int turn = 0;;) {
@@ -565,10 +603,26 @@ __global__ void __launch_bounds__(tc_threads<NH>(), 1)
                 stream_take(js, sj, gj, ct);
                 const int64_t rt = gj;
                 turn = (sj + 1) % NS;
+                int64_t arow0 = rt * BM;
+                if (PK) {  // A comes from the stream's scratch slot of this tile
+                    uint32_t pc = sj == 0 ? pcnt[0] : pcnt[NS - 1];
+                    if ((sj == 0 ? ptile[0] : ptile[NS - 1]) != gj) {  // a new tile: wait for its expansion
+                        if (!mbar_wait(sready_bar(sj, pc & 1u), (pc >> 1) & 1u, abort_flag)) goto producer_done;
+                        ++pc;
+                        if (sj == 0) {
+                            ptile[0] = gj;
+                            pcnt[0] = pc;
+                        } else {
+                            ptile[NS - 1] = gj;
+                            pcnt[NS - 1] = pc;
+                        }
+                    }
+                    arow0 = (((int64_t)blockIdx.x * NS + sj) * 2 + ((pc - 1u) & 1u)) * BM;
+                }
                 {
                     for (int kt = 0; kt < NSEG * p.nkc; ++kt, ++it) {
                         const int seg = kt / p.nkc, kc = kt - seg * p.nkc;
-                        const int arow = (int)(rt * BM) + (NSEG > 1 ? GEMM_SEG_A[seg] * (int)p.n : 0);
+                        const int arow = (int)arow0 + (NSEG > 1 ? GEMM_SEG_A[seg] * (int)p.n : 0);
                         const int brow = ct * BN + (NSEG > 1 ? GEMM_SEG_B[seg] * p.k : 0);
                         const uint32_t s = it % STAGES, ph = (it / STAGES) & 1u;
                         if (!mbar_wait(empty_bar(s), ph ^ 1u, abort_flag)) goto producer_done;
@@ -594,18 +648,41 @@ __global__ void __launch_bounds__(tc_threads<NH>(), 1)
             bool issued = false, gave_up = true;
             uint32_t jc[NS];
             JobStream js[NS];
+            int64_t mtile[NS];  // PK: each stream's current point tile and tiles taken
+            uint32_t mcnt[NS];
             for (int s = 0; s < NS; ++s) {
                 js[s].g = g0 + s * gstep;
                 jc[s] = 0;
+                mtile[s] = -1;
+                mcnt[s] = 0;
                 stream_seek(js[s]);
             }
             for (int turn = 0;; ++job) {
                 const int sj = stream_pick(js, turn);
                 if (sj < 0) break;
+                // PK: whether this job is its tile's last, and the tile's scratch slot
+                bool tile_last = false;
+                uint32_t slot = 0;
                 {
+                    const int hij = sj == 0 ? js[0].hi : js[NS - 1].hi;
                     int64_t gj;
                     int ctj;
                     stream_take(js, sj, gj, ctj);
+                    if (PK) {
+                        uint32_t mc = sj == 0 ? mcnt[0] : mcnt[NS - 1];
+                        if ((sj == 0 ? mtile[0] : mtile[NS - 1]) != gj) {
+                            ++mc;
+                            if (sj == 0) {
+                                mtile[0] = gj;
+                                mcnt[0] = mc;
+                            } else {
+                                mtile[NS - 1] = gj;
+                                mcnt[NS - 1] = mc;
+                            }
+                        }
+                        slot = (mc - 1u) & 1u;
+                        tile_last = ctj == hij - 1;
+                    }
                 }
                 turn = (sj + 1) % NS;
                 {
@@ -619,6 +696,9 @@ __global__ void __launch_bounds__(tc_threads<NH>(), 1)
                     for (int kc = 0; kc < NSEG * p.nkc; ++kc, ++it) {
                         const uint32_t s = it % STAGES, ph = (it / STAGES) & 1u;
                         if (!mbar_wait(full_bar(s), ph, abort_flag)) goto mma_done;
+                        // PK: the tile's last slice has landed, so no TMA load
+                        // reads its scratch slot any more
+                        if (PK && tile_last && kc == NSEG * p.nkc - 1) mbar_arrive(sfree_bar(sj, slot));
                         tc_fence_after();
                         const uint64_t ad = sw128_desc(sA + s * A_STAGE);
                         const uint64_t bd = sw128_desc(sB + s * B_STAGE);
@@ -644,6 +724,78 @@ __global__ void __launch_bounds__(tc_threads<NH>(), 1)
                 mbar_drain(drain_bar, 0u);
             }
         }
+    } else if (PK && warp >= 2 + 4 * NH) {  // -------------------------- converters
+        // Walks the producer's job order and expands a tile at its first job,
+        // ahead of the producer (every tile the producer meets before a tile
+        // this walk waits on has been expanded already, so neither waits on
+        // the other): wait until the stream's scratch slot is free (its tile
+        // two back has had all its A slices loaded), expand the tile's 128
+        // packed rows (bit 1 -> +1.0 = 0x38, bit 0 -> -1.0 = 0xB8, the
+        // tensor-core operand 2 xbar - 1; rows past n as -1) into round16(d)
+        // e4m3 bytes a row, then make the writes visible to the TMA (async
+        // proxy) and mark the slot ready.  Warp w takes rows w, w + CONV_WARPS,
+        // ..., lanes over a row's 32-bit code words; code bits past d meet
+        // zero centroid columns (the B map's width is d).
+        const int cw = warp - (2 + 4 * NH);
+        const int npair = (p.pk_dp + 31) >> 5;  // 32-dimension groups in a scratch row
+        JobStream js[NS];
+        int64_t ctile[NS];
+        uint32_t ccnt[NS];
+        for (int s = 0; s < NS; ++s) {
+            js[s].g = g0 + s * gstep;
+            ctile[s] = -1;
+            ccnt[s] = 0;
+            stream_seek(js[s]);
+        }
+        for (int turn = 0;;) {
+            const int sj = stream_pick(js, turn);
+            if (sj < 0) break;
+            int64_t gj;
+            int ct;
+            stream_take(js, sj, gj, ct);
+            turn = (sj + 1) % NS;
+            if ((sj == 0 ? ctile[0] : ctile[NS - 1]) == gj) continue;  // not a tile's first job
+            const uint32_t i = sj == 0 ? ccnt[0] : ccnt[NS - 1];
+            if (sj == 0) {
+                ctile[0] = gj;
+                ccnt[0] = i + 1;
+            } else {
+                ctile[NS - 1] = gj;
+                ccnt[NS - 1] = i + 1;
+            }
+            const uint32_t slot = i & 1u;
+            if (!mbar_wait(sfree_bar(sj, slot), ((i >> 1) & 1u) ^ 1u, abort_flag)) goto conv_done;
+            // the TMA's reads of the slot's previous tile before these writes
+            asm volatile("fence.proxy.async.global;" ::: "memory");
+            uint8_t *dst = p.pk_scratch + (((size_t)blockIdx.x * NS + sj) * 2 + slot) * BM * p.pk_dp;
+            const int64_t r0 = gj * BM;
+            // lane q takes code word q of the warp's rows (npair <= 32 for
+            // d <= 1024); RB rows' loads in flight before they are expanded
+            const bool act = lane < npair;
+            constexpr int RB = 4;
+            for (int rb = 0; rb < BM / CONV_WARPS; rb += RB) {
+                uint32_t w[RB];
+#pragma unroll
+                for (int u = 0; u < RB; ++u) {
+                    const int64_t row = r0 + cw + CONV_WARPS * (rb + u);
+                    w[u] = act && row < p.n ? __ldg(p.pk_codes + row * p.pk_words + lane) : 0u;
+                }
+#pragma unroll
+                for (int u = 0; u < RB; ++u) {
+                    if (!act) continue;
+                    uint8_t *drow = dst + (size_t)(cw + CONV_WARPS * (rb + u)) * p.pk_dp + 32 * lane;
+                    *reinterpret_cast<uint4 *>(drow) =
+                        make_uint4(pm1_e4m3(w[u]), pm1_e4m3(w[u] >> 4), pm1_e4m3(w[u] >> 8), pm1_e4m3(w[u] >> 12));
+                    if (32 * lane + 16 < p.pk_dp)
+                        *reinterpret_cast<uint4 *>(drow + 16) = make_uint4(
+                            pm1_e4m3(w[u] >> 16), pm1_e4m3(w[u] >> 20), pm1_e4m3(w[u] >> 24), pm1_e4m3(w[u] >> 28));
+                }
+            }
+            asm volatile("fence.proxy.async.global;" ::: "memory");
+            __syncwarp();
+            if (lane == 0) mbar_arrive(sready_bar(sj, slot));
+        }
+    conv_done:;
     } else {  // ------------------------------------------------------- epilogue
         constexpr int NHG = NH / NS;     // warps per TMEM lane quarter in a group
         constexpr int GT = epi_threads<NH>() / NS;  // threads per group
@@ -1552,46 +1704,60 @@ int device_sms() {
     return sms > 0 ? sms : 148;
 }
 
-template <int MODE, bool SEG>
+template <int MODE, bool SEG, bool PK>
 int launch_tc_kind(const void *xs, int64_t n, int dp, int d, const void *cs, int k, const TcParams &p0,
                    cudaStream_t st);
 
+// packed: xs is the 1-bit codes [n][ceil(d/32)] words (MODE_RBQ1 only)
 template <int MODE>
 int launch_tc(const void *xs, int64_t n, int dp, int d, const void *cs, int k, const TcParams &p0,
-              cudaStream_t st) {
-    if (p0.seg_group) return launch_tc_kind<MODE, true>(xs, n, dp, d, cs, k, p0, st);
-    return launch_tc_kind<MODE, false>(xs, n, dp, d, cs, k, p0, st);
+              cudaStream_t st, bool packed = false) {
+    if constexpr (MODE == MODE_RBQ1) {
+        if (packed) {
+            if (p0.seg_group) return launch_tc_kind<MODE, true, true>(xs, n, dp, d, cs, k, p0, st);
+            return launch_tc_kind<MODE, false, true>(xs, n, dp, d, cs, k, p0, st);
+        }
+    }
+    if (p0.seg_group) return launch_tc_kind<MODE, true, false>(xs, n, dp, d, cs, k, p0, st);
+    return launch_tc_kind<MODE, false, false>(xs, n, dp, d, cs, k, p0, st);
 }
 
 // One persistent CTA per SM (at most one point tile per CTA when there are
 // fewer tiles than SMs).
-template <int MODE, bool SEG>
+template <int MODE, bool SEG, bool PK>
 int launch_tc_kind(const void *xs, int64_t n, int dp, int d, const void *cs, int k, const TcParams &p0,
                    cudaStream_t st) {
     constexpr int NH = TC_NH[MODE];
     constexpr int NS = TC_NS[MODE];
     constexpr size_t SMEM = tc_smem_bytes<MODE, NH, NS>();
     static_assert(SMEM <= 227 * 1024, "shared memory per CTA");
-    auto kern = tc_assign_kernel<MODE, NH, SEG, NS>;
-    const int segi = SEG ? 1 : 0;
+    auto kern = tc_assign_kernel<MODE, NH, SEG, NS, PK>;
+    const int segi = SEG ? 1 : 0, pki = PK ? 1 : 0;
     // the dynamic shared memory attribute, set once per device
     constexpr int MAXDEV = 64;
     static std::mutex mu;
-    static bool attr_set[5][2][MAXDEV] = {};
+    static bool attr_set[5][2][2][MAXDEV] = {};
     int dev = 0;
     SKM_CUDA_TRY(cudaGetDevice(&dev));
     {
         std::lock_guard<std::mutex> lock(mu);
-        if (dev >= MAXDEV || !attr_set[MODE][segi][dev]) {
+        if (dev >= MAXDEV || !attr_set[MODE][segi][pki][dev]) {
             SKM_CUDA_TRY(cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)SMEM));
-            if (dev < MAXDEV) attr_set[MODE][segi][dev] = true;
+            if (dev < MAXDEV) attr_set[MODE][segi][pki][dev] = true;
         }
     }
     CUtensorMap ma, mb;
     const int eb = f8_mode<MODE>() ? 1 : 2;
     // GEMM mode: the A and B parts are stacked (rows [part][n], [part][k])
     const int parts = MODE == MODE_GEMM ? 3 : 1;
-    SKM_TRY(make_map(&ma, xs, parts * n, d, dp, BM, eb));
+    // PK: the A slices come from the CTAs' expansion scratch
+    int grid = (int)std::min<int64_t>(device_sms(), cdiv(n, BM));
+    if (PK) {
+        grid = std::min(grid, PK_MAX_CTAS);
+        SKM_TRY(make_map(&ma, p0.pk_scratch, (int64_t)grid * NS * 2 * BM, d, dp, BM, eb));
+    } else {
+        SKM_TRY(make_map(&ma, xs, parts * n, d, dp, BM, eb));
+    }
     SKM_TRY(make_map(&mb, cs, (int64_t)parts * k, d, dp, BN, eb));
     TcParams p = p0;
     p.n = n;
@@ -1600,8 +1766,7 @@ int launch_tc_kind(const void *xs, int64_t n, int dp, int d, const void *cs, int
     p.nct = (int)cdiv(k, BN);
     p.nkc = (int)cdiv(d, 128 / eb);
     p.inject_wait_ns = fault_take(SKM_FAULT_WAIT) ? 1000000ull : 0ull;  // 1 ms
-    const int grid = (int)std::min<int64_t>(device_sms(), p.nrt);
-    kern<<<grid, tc_threads<NH>(), SMEM, st>>>(ma, mb, p);
+    kern<<<grid, tc_threads<NH, PK>(), SMEM, st>>>(ma, mb, p);
     SKM_CUDA_TRY(launched());
     return SKM_OK;
 }
@@ -1614,6 +1779,12 @@ int grid_warps(int64_t items) {
 
 inline int round8(int d) { return (d + 7) & ~7; }
 inline int round16(int d) { return (d + 15) & ~15; }
+// 1-bit codes the tensor-core kernel can read packed (rows a multiple of 16
+// bytes, 16-byte aligned); it does so unless the caller supplies the e4m3
+// screening copy
+inline bool rbq1_packed(int d, const void *x) {
+    return d <= TC_RBQ1_MAX_D && ((d + 31) / 32) % 4 == 0 && ((uintptr_t)x & 15) == 0;
+}
 
 }  // namespace
 
@@ -1656,6 +1827,7 @@ struct ScreenView {
     const float2 *xinfo = nullptr;
     const float *rho_max = nullptr;  // max over points of ||x~ - x|| / ||x~||
     const int32_t *nx = nullptr;
+    bool packed = false;  // RBQ1: xs is the packed codes
 };
 
 static ScreenView screen_view(int repr, int64_t n, int d, const void *x, const void *screen) {
@@ -1681,6 +1853,13 @@ static ScreenView screen_view(int repr, int64_t n, int d, const void *x, const v
         v.rho_max = cv.take<float>(1);
         break;
     case SKM_REPR_RBQ1:
+        if (!screen) {  // no copy: the codes are read packed
+            v.xs = x;
+            v.packed = true;
+            break;
+        }
+        v.xs = cv.take<uint8_t>((size_t)n * round16(d));
+        break;
     case SKM_REPR_LVQ4:
         v.xs = cv.take<uint8_t>((size_t)n * round16(d));
         break;
@@ -1737,7 +1916,8 @@ void tc_plan(int repr, int64_t n, int d, int k, const void *x, const void *scree
                        (repr == SKM_REPR_LVQ4 && d <= TC_LVQ4_MAX_D) ||
                        (repr == SKM_REPR_SQ8 && d <= TC_SQ8_MAX_D);
     if (!dense) return;
-    if (!screen) {
+    const bool pk = repr == SKM_REPR_RBQ1 && !screen && rbq1_packed(d, x);
+    if (!screen && !pk) {
         const size_t sb = tc_screen_bytes(repr, n, d, x);
         b.screen = cv.take<uint8_t>(sb);
     }
@@ -1750,6 +1930,9 @@ void tc_plan(int repr, int64_t n, int d, int k, const void *x, const void *scree
         return;
     }
     if (repr == SKM_REPR_RBQ1) {
+        if (pk)  // read packed: per-CTA expansion slots (two per job stream)
+            b.pk_scratch = cv.take<uint8_t>((size_t)std::min<int64_t>(PK_MAX_CTAS, cdiv(n, BM)) * TC_NS[MODE_RBQ1] *
+                                            2 * BM * round16(d));
         b.cs = reinterpret_cast<uint16_t *>(cv.take<uint8_t>((size_t)k * round16(d)));
         b.rinfo = cv.take<Rbq1CInfo>(k);
         b.rpair_bs = cv.take<float4>(kp / 2);
@@ -1905,7 +2088,8 @@ int tc_assign_rbq1(const skm_data *x, const float *C, int k, int32_t *assign, fl
     const int64_t n = x->n;
     const int d = x->d, dp = round16(d);
     const void *screen = x->screen;
-    if (!screen) {
+    // without a caller copy the codes are read packed where their layout allows
+    if (!screen && !rbq1_packed(d, x->x)) {
         skm_data tmp = *x;
         SKM_TRY(tc_screen_prep(&tmp, b.screen, st));
         screen = b.screen;
@@ -1932,8 +2116,14 @@ int tc_assign_rbq1(const skm_data *x, const float *C, int k, int32_t *assign, fl
     p.F = x->F;
     p.popx = x->popx;
     p.d = d;
+    if (v.packed) {
+        p.pk_codes = static_cast<const uint32_t *>(x->x);
+        p.pk_scratch = b.pk_scratch;
+        p.pk_words = words_of(d);
+        p.pk_dp = dp;
+    }
     SKM_TRY(seg_setup(seg, n, p, st));
-    SKM_TRY(launch_tc<MODE_RBQ1>(v.xs, n, dp, d, b.cs, k, p, st));
+    SKM_TRY(launch_tc<MODE_RBQ1>(v.xs, n, dp, d, b.cs, k, p, st, v.packed));
     add_stats_kernel<<<1, 1, 0, st>>>(b.counters, b.stats);
     SKM_CUDA_TRY(launched());
     return SKM_OK;

@@ -126,7 +126,7 @@ static bool use_prune(const skm_data *x) {
 }
 
 struct AssignBufs {
-    unsigned long long *prune = nullptr;    // [0] pairs alive after block 1, [1] complete
+    unsigned long long *prune = nullptr;    // [0] pairs alive after block 1, [1] complete, [2] later blocks
     int32_t *nx = nullptr, *nc = nullptr;  // SQ8 with d > 1024 (__dp4a path)
     uint4 *planes = nullptr;                // RBQ1 with d > 1024 (AND + popcount path)
     Rbq1CInfo *info = nullptr;
@@ -139,7 +139,7 @@ struct AssignBufs {
 static void plan_assign(const skm_data *x, int k, Carver &cv, AssignBufs &b) {
     const int64_t n = x->n;
     const int d = x->d;
-    b.prune = cv.take<unsigned long long>(2);
+    b.prune = cv.take<unsigned long long>(3);
     if (use_prune(x)) {
         if (x->repr == SKM_REPR_RBQ1) {
             b.planes = cv.take<uint4>((size_t)k * words_of(d));
@@ -751,7 +751,25 @@ int skm_assign(const skm_data *x, const void *C, int k, const int32_t *prev_assi
     AssignBufs b;
     plan_assign(x, k, cv, b);
     SKM_TRY(need_ws(cv, ws_bytes, ws));
+    if (use_prune(x))
+        SKM_CUDA_TRY(cudaMemsetAsync(b.prune, 0, 3 * sizeof(unsigned long long), S(stream)));
     return do_assign(x, C, k, prev_assign, assign, dist, b, S(stream));
+}
+
+int skm_assign_prune_stats(const void *ws, size_t ws_bytes, skm_stats *out, void *stream) {
+    if (!ws || !out) return set_error(SKM_ERR_INVALID_ARG, "ws and out are required");
+    // the counters are the first buffer of every assignment workspace
+    Carver cv(const_cast<void *>(ws), ws_bytes);
+    const unsigned long long *cnt = cv.take<unsigned long long>(3);
+    if (!cv.fits()) return set_error(SKM_ERR_INVALID_ARG, "ws_bytes is smaller than the counters");
+    unsigned long long h[3];
+    SKM_CUDA_TRY(cudaMemcpyAsync(h, cnt, sizeof(h), cudaMemcpyDeviceToHost, S(stream)));
+    SKM_CUDA_TRY(cudaStreamSynchronize(S(stream)));
+    memset(out, 0, sizeof(*out));
+    out->prune_first_block = (int64_t)h[0];
+    out->prune_complete = (int64_t)h[1];
+    out->prune_blocks = (int64_t)h[2];
+    return SKM_OK;
 }
 
 // Segmented assignment (the fine phase of hierarchical k-means): tensor-core
@@ -1119,7 +1137,7 @@ int skm_fit(const skm_fit_config *cfg, const skm_data *x, const void *C_init,
         xd.screen = b.screen;
     }
     SKM_TRY(tc_init_stats(b.a.tc, st));
-    SKM_CUDA_TRY(cudaMemsetAsync(b.a.prune, 0, 2 * sizeof(unsigned long long), st));
+    SKM_CUDA_TRY(cudaMemsetAsync(b.a.prune, 0, 3 * sizeof(unsigned long long), st));
     int e = 0;
     if (x->repr == SKM_REPR_RBQ1) {
         SKM_CUDA_TRY(launch_rbq1_exponent(x->F, n, b.maxbits, b.e_dev, st));
@@ -1202,10 +1220,11 @@ int skm_fit(const skm_fit_config *cfg, const skm_data *x, const void *C_init,
     int32_t uflag = 0;
     SKM_CUDA_TRY(cudaMemcpy(&uflag, b.u.flag, sizeof(uflag), cudaMemcpyDeviceToHost));
     if (uflag) return set_error(SKM_ERR_TIMEOUT, "an update pipeline wait exceeded its limit");
-    unsigned long long pr[2] = {0, 0};
+    unsigned long long pr[3] = {0, 0, 0};
     SKM_CUDA_TRY(cudaMemcpy(pr, b.a.prune, sizeof(pr), cudaMemcpyDeviceToHost));
     local.prune_first_block = (int64_t)pr[0];
     local.prune_complete = (int64_t)pr[1];
+    local.prune_blocks = (int64_t)pr[2];
     if (stats_host) {
         int64_t *per_iter = stats_host->empty_per_iter;
         local.empty_per_iter = per_iter;

@@ -20,6 +20,7 @@ struct TcAssignBufs {
     int64_t *stats = nullptr;     // [0] rescored rows, [1] fallback rows, [2] timeout (cumulative)
     int32_t *counters = nullptr;  // per call: [0] rescore list, [1] fallback list, [2] abort flag
     uint8_t *screen = nullptr;    // screening copy built per call when the caller gave none
+    uint8_t *pk_scratch = nullptr;  // RBQ1 read packed: per-CTA tile expansion slots
     uint16_t *cs = nullptr;       // centroid operand, bf16 [k][round8(d)]
     float4 *cinfo = nullptr;      // F32/BF16: per-column-pair bound terms
     float2 *cinfoz = nullptr;

@@ -86,6 +86,11 @@ def test_invalid_arguments_are_rejected_before_launch(skm):
     assert L.skm_workspace_size(6, ctypes.byref(x8), 32) >= L.skm_workspace_size(7, ctypes.byref(x8), 32) > 0
     # unknown workspace op
     assert L.skm_workspace_size(9, ctypes.byref(x), 4) == 0
+    # pruning counters: no workspace, no output, a workspace too small for them
+    st = skm.Stats()
+    assert L.skm_assign_prune_stats(None, 1 << 20, ctypes.byref(st), None) == 1
+    assert L.skm_assign_prune_stats(FAKE, 1 << 20, None, None) == 1
+    assert L.skm_assign_prune_stats(FAKE, 8, ctypes.byref(st), None) == 1
     # unknown empty-cluster policy
     cfg = skm.FitConfig(4, 3, 7)
     rc = L.skm_fit(ctypes.byref(cfg), ctypes.byref(x), FAKE, None, FAKE, FAKE, None, None, None, FAKE, 1 << 30, None)
@@ -251,3 +256,23 @@ def test_forgy_indices_match_the_oracle(skm):
     assert L.skm_forgy_indices(0, 3, 4, out.ctypes.data) == 1  # k > n
     assert L.skm_forgy_indices(0, 3, 0, out.ctypes.data) == 1
     assert L.skm_forgy_indices(0, 3, 2, None) == 1
+
+
+def test_rbq1_packed_reading_needs_no_screen_workspace(skm):
+    """1-bit rows of a multiple of 16 bytes at a 16-byte aligned address are
+    read packed when no e4m3 screening copy is given, so the assignment
+    workspace holds per-CTA expansion slots instead of a copy of all points;
+    the copy stays available (skm_screen_bytes) for callers who want it."""
+    L = skm.lib()
+
+    def data(d, ptr, n):
+        return skm.Data(2, d, n, ptr, FAKE, FAKE, FAKE, FAKE, 0, 0)
+
+    n = 1_000_000
+    for d in (768, 1024, 100):
+        assert L.skm_screen_bytes(ctypes.byref(data(d, 0x1000, n))) >= n * d
+        packed = L.skm_workspace_size(0, ctypes.byref(data(d, 0x1000, n)), 1000)
+        copied = L.skm_workspace_size(0, ctypes.byref(data(d, 0x1004, n)), 1000)  # misaligned rows
+        assert packed < n * d // 4 and copied >= n * d
+    # 3 words a row: the copy
+    assert L.skm_workspace_size(0, ctypes.byref(data(96, 0x1000, n)), 1000) >= n * 96

@@ -5,6 +5,7 @@ assignments and centroids given identical codes) must be bit-exact; the fp32
 and bf16 paths must agree on >= 99.9% of assignments with every disagreement
 at an oracle top-2 relative gap <= 1e-5, centroids within 1e-4 relative L2
 given identical assignments, objectives within 1e-4 relative."""
+import ctypes
 import math
 
 import numpy as np
@@ -133,6 +134,47 @@ def _skewed_assign(n, k, seed):
     a[torch.rand(n, generator=g) < 0.6] = 0
     a[::997] = -1
     return a
+
+
+def _mixed_size_assign(n, k, seed):
+    """Cluster sizes from {1, 2, 3, 5, 31, 32, 33, 64, 97, 200} in random
+    order (so 32-row chunks of the sorted order hold one, two or many
+    clusters), the rows shuffled, every 501st row outside [0, k)."""
+    g = torch.Generator().manual_seed(seed)
+    choices = torch.tensor([1, 2, 3, 5, 31, 32, 33, 64, 97, 200])
+    sizes = choices[torch.randint(0, len(choices), (k,), generator=g)]
+    lab = torch.repeat_interleave(torch.arange(k, dtype=torch.int32), sizes)
+    lab = torch.cat([lab, torch.randint(0, k, (max(0, n - lab.numel()),), generator=g, dtype=torch.int32)])[:n]
+    a = lab[torch.randperm(n, generator=g)].clone()
+    a[::501] = -1
+    return a
+
+
+@pytest.mark.parametrize("d", [128, 384, 768, 1024])
+@pytest.mark.parametrize("pattern", ["tiny", "mixed"])
+def test_rbq1_update_transposed_table_sums(skm, d, pattern):
+    """The 1-bit fused decode-average sums (bit transposes and subset-sum
+    tables): chunks of 32 sorted rows from one cluster, from two (two table
+    passes), and from many (rows one at a time), ragged last runs and skipped
+    rows, against the oracle bit for bit."""
+    n = 9973
+    if pattern == "tiny":
+        k = 3000
+        a = torch.randint(0, k, (n,), generator=torch.Generator().manual_seed(d), dtype=torch.int32)
+        a[::211] = -1
+    else:
+        k = 150
+        a = _mixed_size_assign(n, k, seed=d + 1)
+    X = _points(n, d, seed=d + 5)
+    r = skm.skm_quantize(skm.REPR_RBQ1, X.to(DEV))
+    pts = skm.rbq1_points(r, d)
+    h = _rbq1_host(r)
+    ok = (a >= 0).numpy()
+    C0 = X[:k].clone()
+    Cn, counts = skm.skm_update(pts, a.to(DEV), C0.to(DEV).clone())
+    Co, co = oracle.rbq1_update(h["codes"][ok], h["F"][ok], d, h["m"], pts.rbq1_exp, a.numpy()[ok], C0.numpy())
+    np.testing.assert_array_equal(counts.cpu().numpy(), co)
+    np.testing.assert_array_equal(Cn.cpu().numpy(), Co)
 
 
 @pytest.mark.parametrize("repr_name,n,d,k", [("f32", 70001, 128, 500), ("f32", 9000, 1536, 40),
@@ -300,7 +342,7 @@ def test_encode_rbq1_vs_oracle(skm, n, d):
 
 
 @pytest.mark.parametrize("n,d,k", [(3000, 768, 300), (777, 33, 7), (500, 64, 1), (1000, 1024, 65),
-                                   (600, 1500, 40)])
+                                   (600, 1500, 40), (2000, 100, 129), (1300, 1000, 300), (257, 128, 513)])
 def test_assign_update_rbq1_bitexact(skm, n, d, k):
     X = _points(n, d, seed=n + 2)
     r = skm.skm_quantize(skm.REPR_RBQ1, X.to(DEV))
@@ -317,6 +359,36 @@ def test_assign_update_rbq1_bitexact(skm, n, d, k):
     Co, co = oracle.rbq1_update(h["codes"], h["F"], d, h["m"], pts.rbq1_exp, ao, C.numpy())
     np.testing.assert_array_equal(counts.cpu().numpy(), co)
     np.testing.assert_array_equal(Cn.cpu().numpy(), Co)
+
+
+@pytest.mark.parametrize("d", [128, 768, 1000])
+def test_assign_rbq1_packed_codes_equal_expanded_copy(skm, d):
+    """Without a screening copy the tensor-core kernel reads 16-byte aligned
+    codes packed (converter warps expand each point tile into a per-CTA slot);
+    with the e4m3 copy, or for misaligned codes, it reads the copy.  All give
+    the oracle's assignment and estimates bit for bit."""
+    n, k = 3001, 260
+    X = _points(n, d, seed=d + 31)
+    r = skm.skm_quantize(skm.REPR_RBQ1, X.to(DEV))
+    pts = skm.rbq1_points(r, d)
+    codes = r["codes"].view(torch.int32).reshape(n, -1)
+    W = codes.shape[1]
+    buf = torch.zeros(n * W + 1, dtype=torch.int32, device=DEV)
+    buf[1:] = codes.reshape(-1)
+    off = buf[1:].view(n, W)  # 4 bytes past a 16-byte boundary
+    assert off.data_ptr() % 16 == 4 and pts.x.data_ptr() % 16 == 0
+    pts_off = skm.Points(skm.REPR_RBQ1, off, d, pts.nx2, pts.F, pts.popx, pts.m, pts.rbq1_exp)
+    C = X[synth.forgy_indices(n, k, seed=3)].clone().to(DEV)
+    a, est = skm.skm_assign(pts, C)
+    a2, est2 = skm.skm_assign(pts_off, C)
+    a3, est3 = skm.skm_assign(pts.with_screen(), C)
+    h = _rbq1_host(r)
+    ao, esto = oracle.rbq1_assign(h["codes"], h["nx2"], h["F"], h["popx"], d,
+                                  oracle.rbq1_centroid_sq4(C.cpu().numpy(), h["m"]))
+    np.testing.assert_array_equal(a.cpu().numpy(), ao)
+    np.testing.assert_array_equal(est.cpu().numpy(), esto)
+    assert torch.equal(a, a2) and torch.equal(est, est2)
+    assert torch.equal(a, a3) and torch.equal(est, est3)
 
 
 def test_fit_rbq1_trajectory_bitexact(skm):
@@ -457,10 +529,21 @@ def test_prune_assign_vs_oracle_and_seed_independent(skm, repr_name, n, d, k):
     _check_f32(a0.cpu().numpy(), d0.cpu().numpy(), best, second, a_or, f"prune {repr_name}")
     # the seed of the bound changes the work, never the result
     prev = torch.randint(0, k, (n,), generator=torch.Generator().manual_seed(7), dtype=torch.int32).to(DEV)
-    a1, d1 = skm.skm_assign(pp, Cd, prev_assign=prev)
-    a2, d2 = skm.skm_assign(pp, Cd, prev_assign=a0.clone())
+    ws = skm.workspace(skm.OP_ASSIGN, pp, k)
+    a1, d1 = skm.skm_assign(pp, Cd, prev_assign=prev, ws=ws)
+    st1 = skm.skm_assign_prune_stats(ws)
+    a2, d2 = skm.skm_assign(pp, Cd, prev_assign=a0.clone(), ws=ws)
+    st2 = skm.skm_assign_prune_stats(ws)  # counters restart with every call
     assert torch.equal(a1, a0) and torch.equal(a2, a0)
     assert torch.equal(d1, d0) and torch.equal(d2, d0)
+    nb = (d + 31) // 32
+    for st in (st1, st2):
+        # every pair evaluates its first block; a pair alive after block b
+        # evaluates block b + 1; complete pairs evaluated all nb blocks
+        assert 0 < st["prune_complete"] <= st["prune_first_block"] <= n * k
+        assert st["prune_complete"] * (nb - 1) <= st["prune_blocks"] <= st["prune_first_block"] * (nb - 1)
+    # the bound from the nearest centroid leaves no more work than a random one
+    assert st2["prune_blocks"] <= st1["prune_blocks"] and st2["prune_first_block"] <= st1["prune_first_block"]
     # and the tensor-core screen reaches the same assignment
     a3, _ = skm.skm_assign(pts, Cd)
     assert (a3 == a0).float().mean().item() >= AGREE
