@@ -233,6 +233,23 @@ def _event_ms(fn, reps, stream):
     return statistics.mean(ts)
 
 
+def _split_ms(fns, reps, stream):
+    """Mean CUDA-event time of each of fns over reps rounds of calling them in
+    order (each bracketed alone)."""
+    import torch
+
+    ts = [[] for _ in fns]
+    for _ in range(reps):
+        for i, fn in enumerate(fns):
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record(stream)
+            fn()
+            e1.record(stream)
+            torch.cuda.synchronize()
+            ts[i].append(e0.elapsed_time(e1))
+    return [statistics.mean(t) for t in ts]
+
+
 def cpu_baseline_c4(Yb_host, C_host, K, budget_s=15.0):
     """Oracle (as it stands) on a bounded row sample of the headline
     workload: one Lloyd iteration (assignment against all k centroids in fp64,
@@ -391,7 +408,9 @@ def run_ours(args):
     # ---- inputs (per-rank shard), resident in HBM before timing -------------
     Yb, C, idx, proj = setup_head(dev, rank, world, dist, peaks)
     N, K = Yb.shape[0], C.shape[0]
-    pts = skm.Points(skm.REPR_BF16, Yb, D_PCA).with_screen()  # per-point norms, built once
+    # per-point norms built once; FLAG_WARM: the same points and assignment
+    # workspace every step, so each screen starts from the previous bounds
+    pts = skm.Points(skm.REPR_BF16, Yb, D_PCA, flags=0 if args.cold_screen else skm.FLAG_WARM).with_screen()
     wsA = skm.workspace(skm.OP_ASSIGN, pts, K)
     wsU = skm.workspace(skm.OP_UPDATE, pts, K)
     a = torch.empty(N, dtype=torch.int32, device=dev)
@@ -417,8 +436,10 @@ def run_ours(args):
     value = world * float(N) * K * args.steps / (ms / 1e3)
 
     # ---- per-kernel times (eager calls after the timed region) ----------------
-    t_assign = _event_ms(lambda: skm.skm_assign(pts, C_step, K, want_dist=False, ws=wsA, out=a), 3, stream)
-    t_update = _event_ms(lambda: skm.skm_update(pts, a, C_step.clone(), counts=cnt, ws=wsU), 3, stream)
+    # assignment and update each timed inside eager steps (every assignment
+    # after an update, as in the timed region)
+    t_assign, t_update = _split_ms([lambda: skm.skm_assign(pts, C_step, K, want_dist=False, ws=wsA, out=a),
+                                    lambda: skm.skm_update(pts, a, C_step, counts=cnt, ws=wsU)], 3, stream)
     long_region = ms > 1000.0
     bf16_peak = peaks["bf16_tflops_sustained"] if long_region else peaks["bf16_tflops"]
     flops = 2.0 * N * K * D_PCA
@@ -1003,6 +1024,8 @@ def main():
                          "assign_rbq1_popcount|assign_prune|assign_prune_sq8|update_f32|update_rbq1|update_sq8|"
                          "update_lvq4|project|quantize_sq8|quantize_rbq1|quantize_lvq4")
     ap.add_argument("--n", type=int, default=200_000)
+    ap.add_argument("--cold-screen", action="store_true",
+                    help="headline step without SKM_FLAG_WARM (every screen starts with no bound)")
     ap.add_argument("--e4m3-copy", action="store_true",
                     help="--case assign_rbq1: read the points from their e4m3 copy instead of packed")
     ap.add_argument("--d", type=int, default=768)

@@ -96,7 +96,20 @@ enum {
      * order), u = fy (d - 2 h), est = fma(-2 F, u, nx2 + ||rho||^2).  Tensor
      * cores (e4m3 +-1 codes on both sides) for d <= 1024, XOR + POPC beyond.
      * The update is unchanged (the points' fused decode-average). */
-    SKM_FLAG_SYMMETRIC = 2
+    SKM_FLAG_SYMMETRIC = 2,
+    /* F32 / BF16 (tensor-core screen) only: the points and the workspace are
+     * those of the previous skm_assign call on this workspace, as between
+     * Lloyd iterations.  Each row decided by the screen leaves in the
+     * workspace an upper bound U on s = ||c||^2 - 2 <x, c> for its centroid;
+     * the next call grows it by that centroid's move (s(x, c') <= U + (||c'||^2
+     * - ||c||^2) + 2 ||x|| ||c' - c||, both terms from the copy of the
+     * previous centroids it keeps) and starts the row's threshold there, so
+     * pairs far from the nearest are not listed as candidates.  The result
+     * is the same; only the work changes.  A workspace whose last call had
+     * other n, d or k, or did not finish, starts cold.  The caller must not
+     * change the points between such calls.  skm_fit uses it between its
+     * iterations. */
+    SKM_FLAG_WARM = 4
 };
 
 /* Points being clustered.  Which fields are read depends on repr. */

@@ -24,7 +24,7 @@ __all__ = [
 ]
 
 REPR_F32, REPR_SQ8, REPR_RBQ1, REPR_BF16, REPR_LVQ4 = 0, 1, 2, 3, 4
-FLAG_PRUNE, FLAG_SYMMETRIC = 1, 2
+FLAG_PRUNE, FLAG_SYMMETRIC, FLAG_WARM = 1, 2, 4
 DTYPE_F32, DTYPE_BF16 = 0, 1
 EMPTY_KEEP, EMPTY_SPLIT = 0, 1
 OP_ASSIGN, OP_UPDATE, OP_FIT, OP_QUANTIZE, OP_PCA, OP_ASSIGN_SEG = 0, 1, 2, 3, 4, 5

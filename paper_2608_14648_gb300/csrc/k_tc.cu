@@ -61,6 +61,8 @@ constexpr int B_STAGE = BN * BK * 2;  // 32 KiB
 // per (point tile, centroid tile) job.
 constexpr int CONV_WARPS = 4;
 constexpr int PK_MAX_CTAS = 160;
+// SKM_FLAG_WARM: stamp word 0 of a workspace whose last call completed
+constexpr int64_t WARM_MAGIC = 0x534b4d5741524d31LL;
 constexpr int TCAND = 4;
 constexpr unsigned long long WAIT_LIMIT_NS = 2000000000ull;  // 2 s per barrier wait
 
@@ -150,6 +152,13 @@ struct TcParams {
     const uint32_t *pk_codes;
     uint8_t *pk_scratch;
     int pk_words, pk_dp;
+    // SCREEN with SKM_FLAG_WARM (NULL otherwise): per row (bits of the bound
+    // U on s for its centroid, that centroid) read at the start and written
+    // at the end; per centroid (||c'||^2 - ||c||^2, ||c' - c||) since the
+    // bounds were written; whether they apply (set by the centroid prep)
+    int2 *warm_row;
+    const float2 *warm_shift;
+    const int32_t *warm_ok;
     // Segmented mode (all NULL otherwise): the point rows are sorted by
     // group and row r may only take centroids [seg_base[g], seg_base[g + 1])
     // of its group g = seg_group[r]; point tile rt covers the centroid tiles
@@ -882,6 +891,22 @@ __global__ void __launch_bounds__(tc_threads<NH, PK>(), 1)
                 a2 = valid ? 2.0f * p.xinfo[row].x : 0.0f;
                 // 2 W_row, W_row = 2 ||x~|| max h' + max z >= every pair's half-width
                 w2 = 2.0f * __fmaf_ru(a2, __ldg(p.hz), __ldg(p.hz + 1));
+                if (p.warm_row && valid && *p.warm_ok) {
+                    // s for the centroid the row had is at most U grown by its move:
+                    // s(x, c') <= U + (||c'||^2 - ||c||^2) + 2 ||x|| ||c' - c||, with
+                    // ||x|| <= ||x~|| + ||x~ - x||.  The nearest centroid j* has
+                    // s~_j* <= s_j* + W_row, so a running minimum started at
+                    // Un - W_row keeps the threshold (minimum + 2 W_row) above it.
+                    const int2 wr = p.warm_row[row];
+                    const float U = __int_as_float(wr.x);
+                    if (wr.y >= 0 && wr.y < p.k && U < INFINITY) {
+                        const float2 sh = __ldg(p.warm_shift + wr.y);
+                        const float2 xi = p.xinfo[row];
+                        const float xn = __fadd_ru(xi.x, xi.y);
+                        const float Un = __fmaf_ru(2.0f * xn, sh.y, __fadd_ru(U, sh.x));
+                        if (Un < INFINITY) sr.umin = __fsub_ru(Un, 0.5f * w2);
+                    }
+                }
             } else if (MODE == MODE_SQ8) {
                 nxr = valid ? p.nx[row] : 0;
             } else if (MODE == MODE_LVQ4) {
@@ -1251,6 +1276,19 @@ __global__ void __launch_bounds__(tc_threads<NH, PK>(), 1)
                     }
                     const int first = kj[0] < p.k ? kj[0] : 0;
                     p.assign[row] = first;
+                    if (p.warm_row) {
+                        // SKM_FLAG_WARM: a decided row keeps U = s~ + W_row >= s for
+                        // its centroid; rows left to the fp32 passes keep none
+                        int2 wr = make_int2(__float_as_int(INFINITY), -1);
+                        if (!overflow && nk == 1) {
+                            float Lj = INFINITY;
+#pragma unroll
+                            for (int t = 0; t < TCAND; ++t)
+                                if (sr.J[t] == kj[0]) Lj = fminf(Lj, sr.L[t]);
+                            wr = make_int2(__float_as_int(__fadd_ru(Lj, 0.5f * w2)), kj[0]);
+                        }
+                        p.warm_row[row] = wr;
+                    }
                     if (!overflow && nk == 1) {
                         // decided by the screen
                     } else if (!overflow && nk >= 2) {
@@ -1396,14 +1434,27 @@ __global__ void screen_prep_sq8_kernel(const uint8_t *__restrict__ X, int64_t n,
 // Records j in [k, kp) get ||c||^2 = +inf so they never matter.  Layout:
 // column pair p = (2p, 2p+1) -> cinfo[p] = (||c||^2 x2, h' x2), cinfoz[p] = (z x2);
 // hz_bits (zeroed by the caller) receives max h' and max z over j < k.
+//
+// SKM_FLAG_WARM (cprev non-NULL): also shift[j] = (||c_j||^2 - ||cprev_j||^2,
+// ||c_j - cprev_j||), each rounded up (fp64 sums of products of fp32 values,
+// plus a margin far above their rounding), then cprev_j = c_j; thread 0
+// publishes in *warm_ok whether the stamp names this n, d and k (the bounds
+// and cprev then belong to these points) and clears the stamp until this
+// call completes.
 __global__ void cprep_f32_kernel(const float *__restrict__ C, int k, int kp, int d, int dp,
                                  float eps_acc, float eps_s, const float *__restrict__ rho_max,
                                  __nv_bfloat16 *__restrict__ cs, float4 *__restrict__ cinfo,
-                                 float2 *__restrict__ cinfoz, unsigned int *__restrict__ hz_bits) {
+                                 float2 *__restrict__ cinfoz, unsigned int *__restrict__ hz_bits,
+                                 float *__restrict__ cprev, float2 *__restrict__ shift,
+                                 int64_t *__restrict__ warm_hdr, int64_t n, int32_t *__restrict__ warm_ok) {
     const int lane = threadIdx.x & 31;
     const int warp = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
     const int nw = (gridDim.x * blockDim.x) >> 5;
     const double rho = (double)*rho_max;
+    if (cprev && blockIdx.x == 0 && threadIdx.x == 0) {
+        *warm_ok = warm_hdr[0] == WARM_MAGIC && warm_hdr[1] == n && warm_hdr[2] == d && warm_hdr[3] == k;
+        warm_hdr[0] = 0;
+    }
     float *cf = reinterpret_cast<float *>(cinfo);
     float *zf = reinterpret_cast<float *>(cinfoz);
     for (int j = warp; j < kp; j += nw) {
@@ -1416,7 +1467,7 @@ __global__ void cprep_f32_kernel(const float *__restrict__ C, int k, int kp, int
             }
             continue;
         }
-        double c2 = 0.0, e2 = 0.0;
+        double c2 = 0.0, e2 = 0.0, p2 = 0.0, dd = 0.0, dn = 0.0;
         for (int i = lane; i < d; i += 32) {
             const float c = C[(int64_t)j * d + i];
             const __nv_bfloat16 cb = __float2bfloat16_rn(c);
@@ -1424,11 +1475,27 @@ __global__ void cprep_f32_kernel(const float *__restrict__ C, int k, int kp, int
             const double cf = (double)__bfloat162float(cb);
             c2 += (double)c * (double)c;
             e2 += (cf - (double)c) * (cf - (double)c);
+            if (cprev) {
+                const double cq = (double)cprev[(int64_t)j * d + i];
+                p2 += cq * cq;
+                dd += ((double)c - cq) * ((double)c - cq);
+                dn += ((double)c - cq) * ((double)c + cq);
+                cprev[(int64_t)j * d + i] = c;
+            }
         }
 #pragma unroll
         for (int o = 16; o > 0; o >>= 1) {
             c2 += __shfl_xor_sync(0xffffffffu, c2, o);
             e2 += __shfl_xor_sync(0xffffffffu, e2, o);
+            if (cprev) {
+                p2 += __shfl_xor_sync(0xffffffffu, p2, o);
+                dd += __shfl_xor_sync(0xffffffffu, dd, o);
+                dn += __shfl_xor_sync(0xffffffffu, dn, o);
+            }
+        }
+        if (cprev && lane == 0) {
+            const double margin = 1e-12 * (c2 + p2);
+            shift[j] = make_float2(__double2float_ru(dn + margin), __double2float_ru(sqrt(dd + margin) * (1.0 + 1e-12)));
         }
         if (lane == 0) {
             const double up = 1.0 + 1e-6;
@@ -1555,13 +1622,24 @@ __device__ __forceinline__ float warp_sqdist(const TX *x, const float *c, int d,
 
 // One warp per listed row: exact fp32 distances to its screen candidates.
 template <typename TX>
+// (count: the call's counters, [0] rows listed, [2] the screen's abort flag.)
+// SKM_FLAG_WARM: thread 0 stamps the workspace's bounds as complete for this
+// n, d and k unless the screen gave up.
 __global__ void rescore_kernel(const TX *__restrict__ X, int d, const float *__restrict__ C,
                                const int32_t *__restrict__ rows, const int32_t *__restrict__ count,
-                               const int32_t *__restrict__ cand, int32_t *__restrict__ assign) {
+                               const int32_t *__restrict__ cand, int32_t *__restrict__ assign,
+                               int64_t *__restrict__ warm_hdr, int64_t n, int k) {
     const int lane = threadIdx.x & 31;
     const int64_t warp = (blockIdx.x * (int64_t)blockDim.x + threadIdx.x) >> 5;
     const int64_t nw = ((int64_t)gridDim.x * blockDim.x) >> 5;
     const int64_t cnt = *count;
+    if (warm_hdr && blockIdx.x == 0 && threadIdx.x == 0 && count[2] == 0) {
+        warm_hdr[1] = n;
+        warm_hdr[2] = d;
+        warm_hdr[3] = k;
+        __threadfence();
+        warm_hdr[0] = WARM_MAGIC;
+    }
     for (int64_t i = warp; i < cnt; i += nw) {
         const int64_t r = rows[i];
         const int32_t *cr = cand + r * (TCAND + 1);
@@ -1905,7 +1983,9 @@ int tc_screen_prep(const skm_data *x, void *screen, cudaStream_t st) {
     return SKM_OK;
 }
 
-void tc_plan(int repr, int64_t n, int d, int k, const void *x, const void *screen, Carver &cv,
+bool tc_rbq1_reads_packed(int d, const void *x) { return rbq1_packed(d, x); }
+
+void tc_plan(int repr, int64_t n, int d, int k, const void *x, const void *screen, bool warm, Carver &cv,
              TcAssignBufs &b) {
     b.stats = cv.take<int64_t>(4);
     b.counters = cv.take<int32_t>(8);  // [4], [5]: SCREEN max h', max z (float bits)
@@ -1943,6 +2023,12 @@ void tc_plan(int repr, int64_t n, int d, int k, const void *x, const void *scree
     if (repr == SKM_REPR_SQ8) {
         b.nc = cv.take<int32_t>(kp);
     } else {
+        if (warm) {
+            b.warm_hdr = cv.take<int64_t>(4);
+            b.warm_row = cv.take<int2>(n);
+            b.warm_cprev = cv.take<float>((size_t)k * d);
+            b.warm_shift = cv.take<float2>(k);
+        }
         b.cinfo = cv.take<float4>(kp / 2);
         b.cinfoz = cv.take<float2>(kp / 2);
         b.cand = cv.take<int32_t>((size_t)n * (TCAND + 1));
@@ -1991,9 +2077,13 @@ int tc_assign_float(const skm_data *x, const float *C, int k, int32_t *assign, f
     const float eps_s = 0x1p-21f;
     const int kp = (int)(cdiv(k, BN) * BN);
     SKM_CUDA_TRY(cudaMemsetAsync(b.counters, 0, sizeof(int32_t) * 8, st));
+    // SKM_FLAG_WARM (not in segmented calls): bounds carried between calls
+    const bool warm = !seg && (x->flags & SKM_FLAG_WARM) && b.warm_hdr;
     cprep_f32_kernel<<<grid_warps(kp), 256, 0, st>>>(C, k, kp, d, dp, eps_acc, eps_s, v.rho_max,
                                                      (__nv_bfloat16 *)b.cs, b.cinfo, b.cinfoz,
-                                                     reinterpret_cast<unsigned int *>(b.counters + 4));
+                                                     reinterpret_cast<unsigned int *>(b.counters + 4),
+                                                     warm ? b.warm_cprev : nullptr, b.warm_shift, b.warm_hdr, n,
+                                                     b.counters + 6);
     SKM_CUDA_TRY(launched());
     TcParams p{};
     p.cinfo = b.cinfo;
@@ -2005,12 +2095,18 @@ int tc_assign_float(const skm_data *x, const float *C, int k, int32_t *assign, f
     p.fall_rows = b.fall_rows;
     p.counters = b.counters;
     p.assign = assign;
+    if (warm) {
+        p.warm_row = b.warm_row;
+        p.warm_shift = b.warm_shift;
+        p.warm_ok = b.counters + 6;
+    }
     SKM_TRY(seg_setup(seg, n, p, st));
     SKM_TRY(launch_tc<MODE_SCREEN>(v.xs, n, dp, d, b.cs, k, p, st));
+    int64_t *hdr = warm ? b.warm_hdr : nullptr;
     const int gw = grid_warps(n);
     if (bf16) {
         const uint16_t *X = static_cast<const uint16_t *>(x->x);
-        rescore_kernel<uint16_t><<<gw, 256, 0, st>>>(X, d, C, b.resc_rows, b.counters, b.cand, assign);
+        rescore_kernel<uint16_t><<<gw, 256, 0, st>>>(X, d, C, b.resc_rows, b.counters, b.cand, assign, hdr, n, k);
         SKM_CUDA_TRY(launched());
         if (seg) {
             seg_rows_exact_kernel<uint16_t><<<gw, 256, 0, st>>>(X, d, C, b.fall_rows, b.counters + 1, seg->group,
@@ -2026,7 +2122,7 @@ int tc_assign_float(const skm_data *x, const float *C, int k, int32_t *assign, f
         }
     } else {
         const float *X = static_cast<const float *>(x->x);
-        rescore_kernel<float><<<gw, 256, 0, st>>>(X, d, C, b.resc_rows, b.counters, b.cand, assign);
+        rescore_kernel<float><<<gw, 256, 0, st>>>(X, d, C, b.resc_rows, b.counters, b.cand, assign, hdr, n, k);
         SKM_CUDA_TRY(launched());
         if (seg) {
             seg_rows_exact_kernel<float><<<gw, 256, 0, st>>>(X, d, C, b.fall_rows, b.counters + 1, seg->group,

@@ -145,7 +145,7 @@ static void plan_assign(const skm_data *x, int k, Carver &cv, AssignBufs &b) {
             b.planes = cv.take<uint4>((size_t)k * words_of(d));
             b.seginfo = cv.take<Rbq1SegInfo>(k);
         }
-        tc_plan(-1, n, d, k, x->x, x->screen, cv, b.tc);  // statistics only
+        tc_plan(-1, n, d, k, x->x, x->screen, false, cv, b.tc);  // statistics only
         return;
     }
     switch (x->repr) {
@@ -170,7 +170,7 @@ static void plan_assign(const skm_data *x, int k, Carver &cv, AssignBufs &b) {
     default:
         break;
     }
-    tc_plan(x->repr, n, d, k, x->x, x->screen, cv, b.tc);
+    tc_plan(x->repr, n, d, k, x->x, x->screen, (x->flags & SKM_FLAG_WARM) != 0, cv, b.tc);
 }
 
 struct UpdateBufs {
@@ -222,7 +222,10 @@ struct FitBufs {
 
 static void plan_fit(const skm_data *x, int k, Carver &cv, FitBufs &b) {
     skm_data xs = *x;
-    if (!x->screen) {
+    if (x->repr == SKM_REPR_F32 || x->repr == SKM_REPR_BF16) xs.flags |= SKM_FLAG_WARM;  // as skm_fit
+    // 1-bit codes the tensor-core kernel reads packed: no copy of the points
+    const bool packed = x->repr == SKM_REPR_RBQ1 && tc_rbq1_reads_packed(x->d, x->x);
+    if (!x->screen && !packed) {
         const size_t sb = tc_screen_bytes(x->repr, x->n, x->d, x->x);
         if (sb) {
             b.screen = cv.take<uint8_t>(sb);
@@ -1136,6 +1139,8 @@ int skm_fit(const skm_fit_config *cfg, const skm_data *x, const void *C_init,
         SKM_TRY(tc_screen_prep(x, b.screen, st));
         xd.screen = b.screen;
     }
+    // the iterations' screens start from the bounds the previous one left
+    if (x->repr == SKM_REPR_F32 || x->repr == SKM_REPR_BF16) xd.flags |= SKM_FLAG_WARM;
     SKM_TRY(tc_init_stats(b.a.tc, st));
     SKM_CUDA_TRY(cudaMemsetAsync(b.a.prune, 0, 3 * sizeof(unsigned long long), st));
     int e = 0;

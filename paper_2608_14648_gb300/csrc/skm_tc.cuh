@@ -21,6 +21,13 @@ struct TcAssignBufs {
     int32_t *counters = nullptr;  // per call: [0] rescore list, [1] fallback list, [2] abort flag
     uint8_t *screen = nullptr;    // screening copy built per call when the caller gave none
     uint8_t *pk_scratch = nullptr;  // RBQ1 read packed: per-CTA tile expansion slots
+    // F32/BF16 with SKM_FLAG_WARM: stamp of the last complete call (magic, n,
+    // d, k), per row (bound bits, centroid), the previous centroids, and per
+    // centroid (||c'||^2 - ||c||^2, ||c' - c||) rounded up
+    int64_t *warm_hdr = nullptr;
+    int2 *warm_row = nullptr;
+    float *warm_cprev = nullptr;
+    float2 *warm_shift = nullptr;
     uint16_t *cs = nullptr;       // centroid operand, bf16 [k][round8(d)]
     float4 *cinfo = nullptr;      // F32/BF16: per-column-pair bound terms
     float2 *cinfoz = nullptr;
@@ -48,7 +55,10 @@ struct TcSeg {
 
 size_t tc_screen_bytes(int repr, int64_t n, int d, const void *x);
 int tc_screen_prep(const skm_data *x, void *screen, cudaStream_t st);
-void tc_plan(int repr, int64_t n, int d, int k, const void *x, const void *screen, Carver &cv,
+// whether the 1-bit tensor-core assignment reads these codes packed when
+// no screening copy is given
+bool tc_rbq1_reads_packed(int d, const void *x);
+void tc_plan(int repr, int64_t n, int d, int k, const void *x, const void *screen, bool warm, Carver &cv,
              TcAssignBufs &b);
 int tc_init_stats(TcAssignBufs &b, cudaStream_t st);
 int tc_assign_float(const skm_data *x, const float *C, int k, int32_t *assign, float *dist,

@@ -549,6 +549,63 @@ def test_prune_assign_vs_oracle_and_seed_independent(skm, repr_name, n, d, k):
     assert (a3 == a0).float().mean().item() >= AGREE
 
 
+@pytest.mark.parametrize("repr_name", ["bf16", "f32"])
+def test_warm_screen_bounds_across_lloyd_steps(skm, repr_name):
+    """SKM_FLAG_WARM: each call starts every row's screen threshold from the
+    bound the previous call left, grown by the centroid's move.  Over Lloyd
+    steps (assign, update) the warm calls give the cold calls' assignment
+    and distances (disagreements only at oracle near-ties) and pass the
+    oracle's checks."""
+    n, d, k, steps = 20011, 256, 300, 4
+    X = _points(n, d, seed=77)
+    if repr_name == "bf16":
+        Xd = X.to(DEV).to(torch.bfloat16).view(torch.int16)
+        xb = Xd.cpu().numpy().view(np.uint16)
+        pts = skm.Points(skm.REPR_BF16, Xd, d)
+        C = torch.from_numpy(oracle.bf16_to_f32(xb[synth.forgy_indices(n, k, seed=6).numpy()]).copy()).to(DEV)
+    else:
+        Xd = X.to(DEV)
+        pts = skm.Points(skm.REPR_F32, Xd, d)
+        C = X[synth.forgy_indices(n, k, seed=6)].clone().to(DEV)
+    warm = pts.with_flags(skm.FLAG_WARM)
+    ws = skm.workspace(skm.OP_ASSIGN, warm, k)
+    for step in range(steps):
+        a_w, d_w = skm.skm_assign(warm, C, ws=ws)
+        a_c, d_c = skm.skm_assign(pts, C)
+        same = (a_w == a_c).float().mean().item()
+        assert same >= 0.9999, f"step {step}: warm and cold agree on {same}"
+        if repr_name == "bf16":
+            a_or, best, second = oracle.assign_bf16(xb, C.cpu().numpy())
+        else:
+            a_or, best, second = oracle.assign_f32(X.numpy(), C.cpu().numpy())
+        _check_f32(a_w.cpu().numpy(), d_w.cpu().numpy(), best, second, a_or, f"warm step {step}")
+        C, _ = skm.skm_update(pts, a_w, C.clone())
+
+
+def test_warm_screen_restarts_cold_on_other_shapes_and_after_abort(skm):
+    """A workspace stamped by a call with another k starts cold; a call that
+    gave up (injected wait) leaves no stamp, so the next warm call starts
+    cold too; every result still equals the cold call's."""
+    n, d = 9000, 128
+    X = _points(n, d, seed=78).to(DEV)
+    pts = skm.Points(skm.REPR_F32, X, d).with_flags(skm.FLAG_WARM)
+    ws = skm.workspace(skm.OP_ASSIGN, pts, 400)
+    C1, C2 = X[:400].clone(), X[1000:1250].clone()
+    skm.skm_assign(pts, C1, ws=ws)
+    a_w, _ = skm.skm_assign(pts, C2, ws=ws)  # k changed: cold
+    a_c, _ = skm.skm_assign(pts.with_flags(0), C2)
+    assert (a_w == a_c).float().mean().item() >= 0.9999
+    skm.skm_assign(pts, C2, ws=ws)  # warm
+    skm.skm_inject_fault(4, 1)  # SKM_FAULT_WAIT: this call's screen gives up before any load
+    skm.skm_assign(pts, (C2 * 1.01).contiguous(), ws=ws)  # asynchronous: its outputs are not used
+    torch.cuda.synchronize()
+    assert skm.skm_fault_armed(4) == 0
+    C3 = (C2 * 0.99).contiguous()
+    a_w, d_w = skm.skm_assign(pts, C3, ws=ws)
+    a_c, d_c = skm.skm_assign(pts.with_flags(0), C3)
+    assert (a_w == a_c).float().mean().item() >= 0.9999
+
+
 def test_prune_fit_bf16(skm):
     n, d, k, iters = 6000, 256, 64, 5
     X = _points(n, d, seed=33)
