@@ -647,6 +647,87 @@ __global__ void __launch_bounds__(RS_THREADS) direct_sum_sq8_kernel(
     cons.finish(lane);
 }
 
+// bf16 rows of at most 1 KB (d <= 512, d % 8 == 0) straight into registers
+// like the SQ8 rows: lane l loads the 16-byte groups l + 32 t (columns
+// 8 (l + 32 t) .. + 7) of a row, a whole row per load instruction of the warp,
+// with the next SQ8_PF rows' loads in flight while one is summed (one bulk
+// copy per 512-byte row left the copy engine, not HBM, as the limit).
+template <typename ACC, int NG>
+__global__ void __launch_bounds__(RS_THREADS) direct_sum_bf16_kernel(
+    const uint16_t *__restrict__ X, int d, const int32_t *__restrict__ perm,
+    const int32_t *__restrict__ scl, const int64_t *__restrict__ offsets, int k, ACC *__restrict__ S,
+    int64_t stride) {
+    __shared__ int32_t sperm_all[RS_CW][RS_ROWS];
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int64_t nval = offsets[k];
+    const int64_t q0 = ((int64_t)blockIdx.x * RS_CW + warp) * RS_ROWS;
+    const int cnt = run_len(nval, q0);
+    if (cnt == 0) return;
+    int32_t *sperm = sperm_all[warp];
+    for (int i = lane; i < cnt; i += 32) sperm[i] = perm[q0 + i];
+    __syncwarp();
+    const int ng = d >> 3;
+    auto load = [&](int r, uint4(&w)[NG]) {
+        const uint4 *src = reinterpret_cast<const uint4 *>(X + (size_t)sperm[r] * d);
+#pragma unroll
+        for (int t = 0; t < NG; ++t)
+            if (lane + 32 * t < ng) w[t] = __ldg(src + lane + 32 * t);
+    };
+    float acc[8 * NG];
+#pragma unroll
+    for (int t = 0; t < 8 * NG; ++t) acc[t] = 0.0f;
+    auto flush = [&](int c) {
+#pragma unroll
+        for (int t = 0; t < NG; ++t)
+#pragma unroll
+            for (int u = 0; u < 8; ++u) {
+                const int col = 8 * (lane + 32 * t) + u;
+                if (col < d) atomicAdd(S + (int64_t)c * stride + col, (ACC)acc[8 * t + u]);
+                acc[8 * t + u] = 0.0f;
+            }
+    };
+    // cluster ids of positions 32 b .. 32 b + 31 (lane-held), this and the next window
+    int clw = lane < cnt ? __ldg(scl + q0 + lane) : -1;
+    int cln = 32 + lane < cnt ? __ldg(scl + q0 + 32 + lane) : -1;
+    int cur = __shfl_sync(0xffffffffu, clw, 0);
+    uint4 buf[SQ8_PF][NG];
+#pragma unroll
+    for (int p = 0; p < SQ8_PF; ++p)
+        if (p < cnt) load(p, buf[p]);
+    for (int r0 = 0; r0 < cnt; r0 += SQ8_PF) {
+#pragma unroll
+        for (int p = 0; p < SQ8_PF; ++p) {
+            const int r = r0 + p;
+            if (r < cnt) {  // warp-uniform
+                if ((r & 31) == 0 && r > 0) {
+                    clw = cln;
+                    const int nx = r + 32 + lane;
+                    cln = nx < cnt ? __ldg(scl + q0 + nx) : -1;
+                }
+                const int c = __shfl_sync(0xffffffffu, clw, r & 31);
+                if (c != cur) {
+                    flush(cur);
+                    cur = c;
+                }
+#pragma unroll
+                for (int t = 0; t < NG; ++t) {
+                    if (lane + 32 * t < ng) {
+                        const uint4 w = buf[p][t];
+                        const uint32_t ww[4] = {w.x, w.y, w.z, w.w};
+#pragma unroll
+                        for (int u = 0; u < 4; ++u) {
+                            acc[8 * t + 2 * u] += __uint_as_float(ww[u] << 16);
+                            acc[8 * t + 2 * u + 1] += __uint_as_float(ww[u] & 0xffff0000u);
+                        }
+                    }
+                }
+                if (r + SQ8_PF < cnt) load(r + SQ8_PF, buf[p]);
+            }
+        }
+    }
+    flush(cur);
+}
+
 // ------------------------------------------------------------- LVQ4 rows
 // T[c][i] += Sq code_i (the fused decode-average of Section 3.1 "LVQ4"),
 // T[c][d] += Bq.  Lane l holds nibble words l + 32 t (t < NW), 8 dimensions
@@ -872,6 +953,19 @@ cudaError_t launch_ring_sum_float(const void *X, int x_is_bf16, int64_t n, int d
                                   const int32_t *scl, const int64_t *offsets, int k, float *S_f,
                                   double *S_d, int32_t *flag, cudaStream_t st) {
     if (n == 0) return cudaSuccess;
+    if (x_is_bf16 && d % 8 == 0 && d <= 512 && (reinterpret_cast<uintptr_t>(X) & 15u) == 0) {
+        // rows of at most 1 KB: straight into registers
+        const unsigned g = ring_blocks(n);
+        const uint16_t *Xb = static_cast<const uint16_t *>(X);
+        if (d <= 256) {
+            if (S_d) direct_sum_bf16_kernel<double, 1><<<g, RS_THREADS, 0, st>>>(Xb, d, perm, scl, offsets, k, S_d, d);
+            else direct_sum_bf16_kernel<float, 1><<<g, RS_THREADS, 0, st>>>(Xb, d, perm, scl, offsets, k, S_f, d);
+        } else {
+            if (S_d) direct_sum_bf16_kernel<double, 2><<<g, RS_THREADS, 0, st>>>(Xb, d, perm, scl, offsets, k, S_d, d);
+            else direct_sum_bf16_kernel<float, 2><<<g, RS_THREADS, 0, st>>>(Xb, d, perm, scl, offsets, k, S_f, d);
+        }
+        return launched();
+    }
     RingLayout L;
     if (!ring_layout((uint32_t)d * (x_is_bf16 ? 2u : 4u), L)) return cudaErrorInvalidValue;
     const int q = (d / 4 + 31) / 32;  // float4 groups per lane

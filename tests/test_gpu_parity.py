@@ -178,7 +178,9 @@ def test_rbq1_update_transposed_table_sums(skm, d, pattern):
 
 
 @pytest.mark.parametrize("repr_name,n,d,k", [("f32", 70001, 128, 500), ("f32", 9000, 1536, 40),
-                                             ("bf16", 20011, 1024, 300), ("rbq1", 70001, 128, 500),
+                                             ("bf16", 20011, 1024, 300), ("bf16", 70001, 256, 500),
+                                             ("bf16", 9001, 200, 40), ("bf16", 20011, 512, 300),
+                                             ("rbq1", 70001, 128, 500),
                                              ("rbq1", 20011, 1024, 300), ("sq8", 70001, 128, 500),
                                              ("sq8", 20011, 1024, 300), ("sq8", 5003, 48, 20)])
 def test_update_skewed_clusters(skm, repr_name, n, d, k):
@@ -464,7 +466,7 @@ def test_pca_fit_vs_oracle(skm):
 
 
 # --------------------------------------------------------- sharded update
-@pytest.mark.parametrize("repr_name", ["f32", "sq8", "rbq1"])
+@pytest.mark.parametrize("repr_name", ["f32", "sq8", "rbq1", "bf16"])
 def test_sharded_update_matches_single(skm, repr_name):
     n, d, k = 4000, 64, 20
     X = _points(n, d, seed=21)
@@ -472,6 +474,11 @@ def test_sharded_update_matches_single(skm, repr_name):
     if repr_name == "f32":
         pts = skm.Points(skm.REPR_F32, Xd, d)
         C = Xd[:k].clone()
+        pdt, pshape = torch.float64, (k, d)
+    elif repr_name == "bf16":  # rows of 128 bytes: the direct register path, fp64 partials
+        Xb = Xd.to(torch.bfloat16).view(torch.int16)
+        pts = skm.Points(skm.REPR_BF16, Xb, d)
+        C = (Xb[:k].to(torch.int32) << 16).view(torch.float32).contiguous()
         pdt, pshape = torch.float64, (k, d)
     elif repr_name == "sq8":
         q = skm.skm_quantize(skm.REPR_SQ8, Xd)
@@ -500,7 +507,7 @@ def test_sharded_update_matches_single(skm, repr_name):
         skm.skm_merge_partials(total, part)
     C_merged = skm.skm_update_finalize(pts, total, counts, C.clone())
     assert torch.equal(counts, cnt_single)
-    if repr_name == "f32":
+    if repr_name in ("f32", "bf16"):
         rel = (C_merged - C_single).norm(dim=1) / C_single.norm(dim=1)
         assert float(rel.max()) <= 1e-5
     else:
