@@ -333,8 +333,8 @@ def run_extra_configs(args, dev, peaks, stream, local_rank):
 
         steps = max(5, min(args.steps, 20))
         ms, launches, timing, clk = _timed_steps(step, stream, steps, 3, 1, None, local_rank, not args.eager)
-        t_a = _event_ms(lambda: skm.skm_assign(pts, C, k, want_dist=False, ws=wsA, out=a), 3, stream)
-        t_u = _event_ms(lambda: skm.skm_update(pts, a, C, counts=cnt, ws=wsU), 3, stream)
+        t_a, t_u = _split_ms([lambda: skm.skm_assign(pts, C, k, want_dist=False, ws=wsA, out=a),
+                              lambda: skm.skm_update(pts, a, C, counts=cnt, ws=wsU)], 3, stream)
         flops = 2.0 * n * k * d
         ach = flops / (t_a / 1e3) / 1e12
         out[name] = {"n": n, "d": d, "k": k, "ms_per_iter": ms / steps, "distances_per_s": n * k * steps / (ms / 1e3),
@@ -354,8 +354,8 @@ def run_extra_configs(args, dev, peaks, stream, local_rank):
     spec = synth.WORKLOADS["emb1m_d768"]
     X = synth.workload_points(spec, seed=0, device=dev)
     idx = synth.forgy_indices(spec.n, spec.k, seed=0).to(dev)
-    timed("emb1m_d768_f32", skm.Points(skm.REPR_F32, X, spec.d).with_screen(), X[idx].clone(), spec.k, spec.n,
-          spec.d, bf16, "bf16")
+    timed("emb1m_d768_f32", skm.Points(skm.REPR_F32, X, spec.d, flags=skm.FLAG_WARM).with_screen(), X[idx].clone(),
+          spec.k, spec.n, spec.d, bf16, "bf16")
     pR = skm.rbq1_points(skm.skm_quantize(skm.REPR_RBQ1, X), spec.d)
     CR, _, _, _, _ = skm.skm_fit(pR, spec.k, 0, init_idx=idx, want_objective=False, want_dist=False)
     timed("emb1m_d768_rbq1", pR, CR, spec.k, spec.n, spec.d, 2 * bf16, "e4m3", copy_pts=pR.with_screen())
