@@ -607,7 +607,15 @@ typedef struct skm_step_host_config {
     int64_t *counts;
     skm_exchange_fn exchange;
     void *user;
-    int32_t reserved[4];
+    int32_t warm;           /* F32 / BF16: 1 when x's host points are those of
+                               the previous call with this workspace and
+                               configuration (Lloyd iterations): each range
+                               keeps its own assignment workspace and its
+                               screen starts from the bounds that range's
+                               previous call left (SKM_FLAG_WARM); the
+                               workspace then holds one assignment workspace
+                               per range.  0: every call starts cold.        */
+    int32_t reserved[3];
 } skm_step_host_config;
 
 size_t skm_step_host_workspace_size(const skm_step_host_config *cfg, const skm_data *x);

@@ -101,7 +101,7 @@ class StepHostConfig(ctypes.Structure):
 
     _fields_ = [("k", ctypes.c_int32), ("chunks", ctypes.c_int32), ("copy_stream", ctypes.c_void_p),
                 ("partial", ctypes.c_void_p), ("counts", ctypes.c_void_p), ("exchange", EXCHANGE_FN),
-                ("user", ctypes.c_void_p), ("reserved", ctypes.c_int32 * 4)]
+                ("user", ctypes.c_void_p), ("warm", ctypes.c_int32), ("reserved", ctypes.c_int32 * 3)]
 
 
 def lib_path() -> str:
@@ -571,9 +571,11 @@ class LloydStepHost:
     held in (pinned) host memory per call.  `exchange` (optional) is a
     callable run between the partial sums and the finalisation; it must
     enqueue its work on the step's stream and then reads/writes the tensors
-    `self.partial` and `self.counts`."""
+    `self.partial` and `self.counts`.  warm=True: the host points do not
+    change between calls, so each row range's screen starts from the bounds
+    its previous call left (one assignment workspace per range)."""
 
-    def __init__(self, repr_, X_host, d, k, chunks=16, device=None, copy_stream=None, exchange=None):
+    def __init__(self, repr_, X_host, d, k, chunks=16, device=None, copy_stream=None, exchange=None, warm=False):
         self.device = torch.device("cuda") if device is None else torch.device(device)
         self.repr, self.k, self.d = repr_, int(k), int(d)
         self.X_host = X_host
@@ -585,7 +587,7 @@ class LloydStepHost:
         self._user_exchange = exchange
         self._cb = EXCHANGE_FN(self._exchange) if exchange is not None else EXCHANGE_FN()
         self.cfg = StepHostConfig(self.k, int(chunks), ctypes.c_void_p(self.copy_stream.cuda_stream),
-                                  self.partial.data_ptr(), self.counts.data_ptr(), self._cb, None)
+                                  self.partial.data_ptr(), self.counts.data_ptr(), self._cb, None, int(bool(warm)))
         nbytes = lib().skm_step_host_workspace_size(ctypes.byref(self.cfg), ctypes.byref(self.ref))
         if nbytes == 0:
             raise SkmError(1, lib().skm_last_error().decode())

@@ -66,7 +66,12 @@ struct HostBufs {
     double *red = nullptr, *chunk_sum = nullptr, *total = nullptr;
     uint8_t *ws_a = nullptr, *ws_u = nullptr;
     size_t ws_a_bytes = 0, ws_u_bytes = 0;
+    size_t ws_a_stride = 0;  // warm: range i's assignment workspace at ws_a + i * ws_a_stride
 };
+
+bool host_warm(const skm_step_host_config *cfg, const skm_data *x) {
+    return cfg->warm && (x->repr == SKM_REPR_F32 || x->repr == SKM_REPR_BF16);
+}
 
 void plan_host(const skm_step_host_config *cfg, const skm_data *x, Carver &cv, HostBufs &b) {
     const int64_t rc = cdiv(x->n, cfg->chunks);
@@ -87,9 +92,13 @@ void plan_host(const skm_step_host_config *cfg, const skm_data *x, Carver &cv, H
     // the entry points' own workspaces for a range of rc rows (reused by
     // every range: the compute stream runs them one after another)
     skm_data probe = view_of(x, reinterpret_cast<const void *>(256), rc);
+    if (host_warm(cfg, x)) probe.flags |= SKM_FLAG_WARM;
     b.ws_a_bytes = skm_workspace_size(0, &probe, k);
+    probe.flags = 0;
     b.ws_u_bytes = skm_workspace_size(1, &probe, k);
-    b.ws_a = cv.take<uint8_t>(b.ws_a_bytes);
+    // warm: one assignment workspace per range (each keeps its rows' bounds)
+    b.ws_a_stride = (b.ws_a_bytes + 255) & ~size_t(255);
+    b.ws_a = cv.take<uint8_t>(host_warm(cfg, x) ? b.ws_a_stride * (size_t)cfg->chunks : b.ws_a_bytes);
     b.ws_u = cv.take<uint8_t>(b.ws_u_bytes);
 }
 
@@ -143,6 +152,7 @@ extern "C" int skm_lloyd_step_host(const skm_step_host_config *cfg, const skm_da
     int64_t *counts = cfg->counts ? cfg->counts : b.counts;
     const size_t cbytes = (size_t)k * d * (x->repr == SKM_REPR_SQ8 ? 1 : 4);
     const char *xh = static_cast<const char *>(x->x);
+    const bool warm = host_warm(cfg, x);
 
     cudaEvent_t landed[RING], freed[RING];
     int made = 0;
@@ -177,9 +187,15 @@ extern "C" int skm_lloyd_step_host(const skm_step_host_config *cfg, const skm_da
             SKM_CUDA_TRY(cudaMemcpyAsync(b.ring[s], xh + r0 * rb, (size_t)(rows * rb), cudaMemcpyHostToDevice, cp));
             SKM_CUDA_TRY(cudaEventRecord(landed[s], cp));
             SKM_CUDA_TRY(cudaStreamWaitEvent(st, landed[s], 0));
-            const skm_data v = view_of(x, b.ring[s], rows);
-            SKM_TRY(skm_assign(&v, b.C, k, nullptr, b.assign[s], objective_host ? b.dist[s] : nullptr, b.ws_a,
+            skm_data v = view_of(x, b.ring[s], rows);
+            uint8_t *wsa = b.ws_a;
+            if (warm) {  // this range's own workspace: its rows' bounds from the previous call
+                v.flags |= SKM_FLAG_WARM;
+                wsa = b.ws_a + (size_t)i * b.ws_a_stride;
+            }
+            SKM_TRY(skm_assign(&v, b.C, k, nullptr, b.assign[s], objective_host ? b.dist[s] : nullptr, wsa,
                                b.ws_a_bytes, st));
+            v.flags = 0;
             SKM_TRY(skm_update(&v, b.assign[s], k, nullptr, counts, partial, b.ws_u, b.ws_u_bytes, st));
             if (objective_host) {
                 const int nblk = (int)std::min<int64_t>(RED, rows);

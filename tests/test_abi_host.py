@@ -180,6 +180,14 @@ def test_step_host_arguments_are_rejected_before_any_work(skm):
         return skm.StepHostConfig(k, chunks, None, None, None, skm.EXCHANGE_FN(), None)
 
     assert L.skm_step_host_workspace_size(ctypes.byref(cfg()), ctypes.byref(x)) > 0
+    # warm: one assignment workspace per range for F32/BF16, nothing extra for SQ8
+    warm = cfg()
+    warm.warm = 1
+    assert L.skm_step_host_workspace_size(ctypes.byref(warm), ctypes.byref(x)) > \
+        L.skm_step_host_workspace_size(ctypes.byref(cfg()), ctypes.byref(x))
+    x8 = skm.Data(1, 16, 100, X.ctypes.data, None, None, None, None, 0, 0)
+    assert L.skm_step_host_workspace_size(ctypes.byref(warm), ctypes.byref(x8)) == \
+        L.skm_step_host_workspace_size(ctypes.byref(cfg()), ctypes.byref(x8))
     for c, code, what in [(cfg(k=101), 1, b"k = 101"), (cfg(k=0), 1, b"k = 0"), (cfg(chunks=0), 1, b"chunks"),
                           (cfg(chunks=257), 1, b"chunks")]:
         assert L.skm_step_host_workspace_size(ctypes.byref(c), ctypes.byref(x)) == 0

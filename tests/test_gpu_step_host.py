@@ -120,3 +120,25 @@ def test_step_host_rejects_pageable_points(skm):
     with pytest.raises(skm.SkmError) as ei:
         step(C0.clone())
     assert ei.value.code == 1
+
+
+@pytest.mark.parametrize("kind,chunks", [("bf16", 16), ("f32", 5)])
+def test_step_host_warm_ranges_match_cold(skm, kind, chunks):
+    """warm=1: each row range keeps its own assignment workspace and starts
+    its screen from the bounds its previous call left.  Over Lloyd
+    iterations (each call's output centroids fed to the next) the warm steps
+    give the cold steps' assignments (near-ties aside) and centroids."""
+    n, d, k = 30011, 128, 200
+    repr_, Xh, C0 = _inputs(skm, kind, n, d, k, seed=41)
+    Xp = Xh.pin_memory()
+    cold = skm.LloydStepHost(repr_, Xp, d, k, chunks=chunks)
+    warm = skm.LloydStepHost(repr_, Xp, d, k, chunks=chunks, warm=True)
+    assert warm.ws.numel() > cold.ws.numel()
+    Cc, Cw = C0.clone().pin_memory(), C0.clone().pin_memory()
+    for it in range(4):
+        _, a_c, _, _ = cold(Cc, Cc)
+        _, a_w, _, _ = warm(Cw, Cw)
+        agree = (a_c == a_w).float().mean().item()
+        assert agree >= 0.9999, f"iteration {it}: agreement {agree}"
+        if agree == 1.0:
+            _close_l2(Cw, Cc)
