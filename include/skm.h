@@ -464,12 +464,11 @@ int skm_assign_prune_stats(const void *ws, size_t ws_bytes, skm_stats *out, void
  * library keeps until exit.
  *   Limits: k <= 16384 and k * ceil(d/32) <= 131072, else SKM_ERR_UNSUPPORTED
  *   (nothing is launched).
- *   The first call on a device looks up the array's device address with that
- *   device current (cudaGetSymbolAddress) and caches it; make that first call
- *   before any stream capture.  The cached address belongs to the device's
- *   current (primary) context: do not use this entry point across a
- *   cudaDeviceReset or anything else that destroys and recreates that context,
- *   because the array then moves and the cached address goes stale.
+ *   Every call looks up the array's device address in the current context
+ *   (cudaGetSymbolAddress, which allocates nothing), so the entry point stays
+ *   valid when that context is destroyed and recreated (cudaDeviceReset); the
+ *   first call on a device may load the library's module, so make it before
+ *   any stream capture.
  *   All calls share the array and it keeps the last call's contents: calls
  *   whose work overlaps on the GPU (other streams, other threads) race; order
  *   them on one stream or synchronise between them.

@@ -11,8 +11,6 @@
 // the per-centroid estimator terms (k records of 16 bytes), the same data
 // skm_assign builds in its workspace.  It lives in one file-scope device array
 // of 2.25 MiB that every GPU which loads the library keeps until exit.
-#include <mutex>
-
 #include "skm_internal.cuh"
 
 namespace skm {
@@ -24,28 +22,15 @@ constexpr size_t NOALLOC_BYTES = NOALLOC_PLANE_WORDS * sizeof(uint4) + NOALLOC_M
 
 static __device__ __align__(256) unsigned char g_rbq1_scratch[NOALLOC_BYTES];
 
-constexpr int MAX_DEVICES = 64;
-std::mutex g_mu;
-void *g_addr[MAX_DEVICES] = {};
-
-// Device address of g_rbq1_scratch on the current device.  The host-side
-// symbol is only a stand-in, so the address is looked up once per device
-// (with that device current) and cached.
+// Device address of g_rbq1_scratch in the current context, looked up on
+// every call (cudaGetSymbolAddress allocates nothing), so the address stays
+// right after the context is torn down and the module loaded again.
 int scratch_address(void **out) {
-    int dev = 0;
-    SKM_CUDA_TRY(cudaGetDevice(&dev));
-    if (dev < 0 || dev >= MAX_DEVICES)
-        return set_error(SKM_ERR_UNSUPPORTED, "device ordinal %d beyond %d", dev, MAX_DEVICES);
-    std::lock_guard<std::mutex> lock(g_mu);
-    if (!g_addr[dev]) {
-        void *p = nullptr;
-        const cudaError_t e = cudaGetSymbolAddress(&p, g_rbq1_scratch);
-        if (e != cudaSuccess || !p)
-            return set_error(SKM_ERR_CUDA, "cudaGetSymbolAddress(g_rbq1_scratch) failed: %s",
-                             cudaGetErrorString(e));
-        g_addr[dev] = p;
-    }
-    *out = g_addr[dev];
+    void *p = nullptr;
+    const cudaError_t e = cudaGetSymbolAddress(&p, g_rbq1_scratch);
+    if (e != cudaSuccess || !p)
+        return set_error(SKM_ERR_CUDA, "cudaGetSymbolAddress(g_rbq1_scratch) failed: %s", cudaGetErrorString(e));
+    *out = p;
     return SKM_OK;
 }
 
