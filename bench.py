@@ -685,7 +685,7 @@ def run_case(args):
         pts = skm.rbq1_points(q, d).with_segments(skm.skm_rbq1_segments(X, q["m"])).with_flags(skm.FLAG_PRUNE)
     elif args.case in ("assign_lvq4", "update_lvq4"):
         pts = skm.lvq4_points(skm.skm_quantize(skm.REPR_LVQ4, X), d)
-        if args.case == "assign_lvq4":
+        if args.case == "assign_lvq4" and args.e4m3_copy:  # the e4m3 screening copy instead of packed codes
             pts = pts.with_screen()
     elif args.case in ("assign_sq8", "update_sq8"):
         q = skm.skm_quantize(skm.REPR_SQ8, X)
@@ -1029,7 +1029,7 @@ def main():
     ap.add_argument("--cold-screen", action="store_true",
                     help="headline step without SKM_FLAG_WARM (every screen starts with no bound)")
     ap.add_argument("--e4m3-copy", action="store_true",
-                    help="--case assign_rbq1: read the points from their e4m3 copy instead of packed")
+                    help="--case assign_rbq1 / assign_lvq4: read the points from their e4m3 copy instead of packed")
     ap.add_argument("--d", type=int, default=768)
     ap.add_argument("--k", type=int, default=1000)
     ap.add_argument("--reps", type=int, default=3)

@@ -387,14 +387,15 @@ int skm_lvq4_exponent(const float *lvq, int64_t n, int *e_host, void *ws, size_t
  * representation needs none: SQ8, RBQ1 or LVQ4 with d > 1024);
  * skm_screen_prep fills `screen` (device, 256-byte aligned,
  * caller-owned) from x->x.  Asynchronous.
- * RBQ1 without a copy (x->screen NULL): when a code row is a multiple of 16
- * bytes (ceil(d/32) a multiple of 4) at a 16-byte aligned address, the
- * assignment reads the codes packed (each CTA expands its point tiles into a
- * slot of the workspace, at most 160 x 4 x 128 x round16(d) bytes), so the
- * points occupy ceil(d/32) words in HBM instead of round16(d) bytes; the copy
- * saves that per-tile expansion (measured on GB300: 1M x 768, k = 1000: 0.61
- * ms packed, 0.53 ms from the copy).  Otherwise skm_assign builds the copy in
- * its workspace on every call. */
+ * RBQ1 / LVQ4 without a copy (x->screen NULL): when a code row is a multiple
+ * of 16 bytes (ceil(d/32), resp. ceil(d/8), a multiple of 4) at a 16-byte
+ * aligned address, the assignment reads the codes packed (each CTA expands
+ * its point tiles into a slot of the workspace, at most 160 x 4 x 128 x
+ * round16(d) bytes), so the points occupy their code words in HBM instead of
+ * round16(d) bytes; the copy saves that per-tile expansion (measured on
+ * GB300, 1M x 768, k = 1000: RBQ1 0.61 ms packed, 0.50 ms from the copy;
+ * LVQ4 0.76 and 0.52 ms; at k = 3162 and d = 1024 the gap is 7-9%).
+ * Otherwise skm_assign builds the copy in its workspace on every call. */
 size_t skm_screen_bytes(const skm_data *x);
 int skm_screen_prep(const skm_data *x, void *screen, size_t screen_bytes, void *stream);
 

@@ -116,9 +116,13 @@ constexpr int REC_BYTES = 4096;
 // merge buffer (per group, slices 1..NH/NS-1 publish) and the record buffers
 // (two per group).
 template <int MODE, int NH, int NS>
+constexpr size_t tc_lut_offset() {  // LVQ4 read packed: byte -> two e4m3 codes, after the records
+    return (size_t)STAGES * (A_STAGE + B_STAGE) + 512 + (size_t)(NH - NS) * BM * merge_words<MODE>() * 4 +
+           2 * NS * REC_BYTES;
+}
+template <int MODE, int NH, int NS>
 constexpr size_t tc_smem_bytes() {
-    return 1024 + (size_t)STAGES * (A_STAGE + B_STAGE) + 512 +
-           (size_t)(NH - NS) * BM * merge_words<MODE>() * 4 + 2 * NS * REC_BYTES;
+    return 1024 + tc_lut_offset<MODE, NH, NS>() + (MODE == 3 /* MODE_LVQ4 */ ? 512 : 0);
 }
 
 struct TcParams {
@@ -500,7 +504,12 @@ __global__ void __launch_bounds__(tc_threads<NH, PK>(), 1)
     // from it has landed)
     auto sready_bar = [&](int j, int i) { return bar0 + 8u * (2 * STAGES + 7 + 2 * j + i); };
     auto sfree_bar = [&](int j, int i) { return bar0 + 8u * (2 * STAGES + 11 + 2 * j + i); };
-    static_assert(!PK || MODE == MODE_RBQ1, "packed points: 1-bit codes only");
+    static_assert(!PK || MODE == MODE_RBQ1 || MODE == MODE_LVQ4, "packed points: 1-bit or LVQ4 codes");
+    // PK, LVQ4: lut[b] = e4m3 codes of the two nibbles of byte b (low byte: low nibble)
+    uint16_t *lut = reinterpret_cast<uint16_t *>(smem + tc_lut_offset<MODE, NH, NS>());
+    if (PK && MODE == MODE_LVQ4)
+        for (int i = threadIdx.x; i < 256; i += blockDim.x)
+            lut[i] = (uint16_t)(e4m3_of_code(i & 15) | ((uint32_t)e4m3_of_code(i >> 4) << 8));
     // the epilogue's merge buffer starts 256 bytes after tmem_slot (see tc_smem_bytes)
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -740,7 +749,8 @@ __global__ void __launch_bounds__(tc_threads<NH, PK>(), 1)
         // the other): wait until the stream's scratch slot is free (its tile
         // two back has had all its A slices loaded), expand the tile's 128
         // packed rows (bit 1 -> +1.0 = 0x38, bit 0 -> -1.0 = 0xB8, the
-        // tensor-core operand 2 xbar - 1; rows past n as -1) into round16(d)
+        // tensor-core operand 2 xbar - 1; rows past n as -1; LVQ4 nibbles ->
+        // their e4m3 integer codes, rows past n as 0) into round16(d)
         // e4m3 bytes a row, then make the writes visible to the TMA (async
         // proxy) and mark the slot ready.  Warp w takes rows w, w + CONV_WARPS,
         // ..., lanes over a row's 32-bit code words; code bits past d meet
@@ -778,26 +788,59 @@ __global__ void __launch_bounds__(tc_threads<NH, PK>(), 1)
             asm volatile("fence.proxy.async.global;" ::: "memory");
             uint8_t *dst = p.pk_scratch + (((size_t)blockIdx.x * NS + sj) * 2 + slot) * BM * p.pk_dp;
             const int64_t r0 = gj * BM;
-            // lane q takes code word q of the warp's rows (npair <= 32 for
-            // d <= 1024); RB rows' loads in flight before they are expanded
-            const bool act = lane < npair;
             constexpr int RB = 4;
-            for (int rb = 0; rb < BM / CONV_WARPS; rb += RB) {
-                uint32_t w[RB];
+            if constexpr (MODE == MODE_RBQ1) {
+                // lane q takes code word q of the warp's rows (npair <= 32 for
+                // d <= 1024); RB rows' loads in flight before they are expanded
+                const bool act = lane < npair;
+                for (int rb = 0; rb < BM / CONV_WARPS; rb += RB) {
+                    uint32_t w[RB];
 #pragma unroll
-                for (int u = 0; u < RB; ++u) {
-                    const int64_t row = r0 + cw + CONV_WARPS * (rb + u);
-                    w[u] = act && row < p.n ? __ldg(p.pk_codes + row * p.pk_words + lane) : 0u;
+                    for (int u = 0; u < RB; ++u) {
+                        const int64_t row = r0 + cw + CONV_WARPS * (rb + u);
+                        w[u] = act && row < p.n ? __ldg(p.pk_codes + row * p.pk_words + lane) : 0u;
+                    }
+#pragma unroll
+                    for (int u = 0; u < RB; ++u) {
+                        if (!act) continue;
+                        uint8_t *drow = dst + (size_t)(cw + CONV_WARPS * (rb + u)) * p.pk_dp + 32 * lane;
+                        *reinterpret_cast<uint4 *>(drow) =
+                            make_uint4(pm1_e4m3(w[u]), pm1_e4m3(w[u] >> 4), pm1_e4m3(w[u] >> 8), pm1_e4m3(w[u] >> 12));
+                        if (32 * lane + 16 < p.pk_dp)
+                            *reinterpret_cast<uint4 *>(drow + 16) = make_uint4(
+                                pm1_e4m3(w[u] >> 16), pm1_e4m3(w[u] >> 20), pm1_e4m3(w[u] >> 24), pm1_e4m3(w[u] >> 28));
+                    }
                 }
+            } else {
+                // LVQ4: lane q takes nibble words q + 32 t (8 dimensions each; at
+                // most 128 words for d <= 1024) of the warp's rows, RB rows' loads
+                // in flight, each byte looked up as two e4m3 codes
+                const int nq = p.pk_dp >> 3;  // 8-dimension words in a scratch row (<= pk_words)
+                for (int rb = 0; rb < BM / CONV_WARPS; rb += RB) {
+                    uint32_t w[RB][4];
 #pragma unroll
-                for (int u = 0; u < RB; ++u) {
-                    if (!act) continue;
-                    uint8_t *drow = dst + (size_t)(cw + CONV_WARPS * (rb + u)) * p.pk_dp + 32 * lane;
-                    *reinterpret_cast<uint4 *>(drow) =
-                        make_uint4(pm1_e4m3(w[u]), pm1_e4m3(w[u] >> 4), pm1_e4m3(w[u] >> 8), pm1_e4m3(w[u] >> 12));
-                    if (32 * lane + 16 < p.pk_dp)
-                        *reinterpret_cast<uint4 *>(drow + 16) = make_uint4(
-                            pm1_e4m3(w[u] >> 16), pm1_e4m3(w[u] >> 20), pm1_e4m3(w[u] >> 24), pm1_e4m3(w[u] >> 28));
+                    for (int u = 0; u < RB; ++u) {
+                        const int64_t row = r0 + cw + CONV_WARPS * (rb + u);
+#pragma unroll
+                        for (int t = 0; t < 4; ++t) {
+                            const int q = lane + 32 * t;
+                            w[u][t] = q < nq && row < p.n ? __ldg(p.pk_codes + row * p.pk_words + q) : 0u;
+                        }
+                    }
+#pragma unroll
+                    for (int u = 0; u < RB; ++u) {
+                        uint8_t *drow = dst + (size_t)(cw + CONV_WARPS * (rb + u)) * p.pk_dp;
+#pragma unroll
+                        for (int t = 0; t < 4; ++t) {
+                            const int q = lane + 32 * t;
+                            if (q < nq) {
+                                const uint32_t v = w[u][t];
+                                *reinterpret_cast<uint2 *>(drow + 8 * q) =
+                                    make_uint2((uint32_t)lut[v & 255u] | ((uint32_t)lut[(v >> 8) & 255u] << 16),
+                                               (uint32_t)lut[(v >> 16) & 255u] | ((uint32_t)lut[v >> 24] << 16));
+                            }
+                        }
+                    }
                 }
             }
             asm volatile("fence.proxy.async.global;" ::: "memory");
@@ -1786,11 +1829,12 @@ template <int MODE, bool SEG, bool PK>
 int launch_tc_kind(const void *xs, int64_t n, int dp, int d, const void *cs, int k, const TcParams &p0,
                    cudaStream_t st);
 
-// packed: xs is the 1-bit codes [n][ceil(d/32)] words (MODE_RBQ1 only)
+// packed: xs is the 1-bit codes [n][ceil(d/32)] or the LVQ4 nibble words
+// [n][ceil(d/8)] (MODE_RBQ1 / MODE_LVQ4)
 template <int MODE>
 int launch_tc(const void *xs, int64_t n, int dp, int d, const void *cs, int k, const TcParams &p0,
               cudaStream_t st, bool packed = false) {
-    if constexpr (MODE == MODE_RBQ1) {
+    if constexpr (MODE == MODE_RBQ1 || MODE == MODE_LVQ4) {
         if (packed) {
             if (p0.seg_group) return launch_tc_kind<MODE, true, true>(xs, n, dp, d, cs, k, p0, st);
             return launch_tc_kind<MODE, false, true>(xs, n, dp, d, cs, k, p0, st);
@@ -1862,6 +1906,11 @@ inline int round16(int d) { return (d + 15) & ~15; }
 // screening copy
 inline bool rbq1_packed(int d, const void *x) {
     return d <= TC_RBQ1_MAX_D && ((d + 31) / 32) % 4 == 0 && ((uintptr_t)x & 15) == 0;
+}
+// the same for LVQ4 nibble words (then round16(d) <= 8 ceil(d/8): every word
+// a converter reads lies inside the row)
+inline bool lvq4_packed(int d, const void *x) {
+    return d <= TC_LVQ4_MAX_D && ((d + 7) / 8) % 4 == 0 && ((uintptr_t)x & 15) == 0;
 }
 
 }  // namespace
@@ -1939,6 +1988,11 @@ static ScreenView screen_view(int repr, int64_t n, int d, const void *x, const v
         v.xs = cv.take<uint8_t>((size_t)n * round16(d));
         break;
     case SKM_REPR_LVQ4:
+        if (!screen) {  // no copy: the codes are read packed
+            v.xs = x;
+            v.packed = true;
+            break;
+        }
         v.xs = cv.take<uint8_t>((size_t)n * round16(d));
         break;
     }
@@ -1983,7 +2037,9 @@ int tc_screen_prep(const skm_data *x, void *screen, cudaStream_t st) {
     return SKM_OK;
 }
 
-bool tc_rbq1_reads_packed(int d, const void *x) { return rbq1_packed(d, x); }
+bool tc_reads_packed(int repr, int d, const void *x) {
+    return (repr == SKM_REPR_RBQ1 && rbq1_packed(d, x)) || (repr == SKM_REPR_LVQ4 && lvq4_packed(d, x));
+}
 
 void tc_plan(int repr, int64_t n, int d, int k, const void *x, const void *screen, bool warm, Carver &cv,
              TcAssignBufs &b) {
@@ -1996,13 +2052,17 @@ void tc_plan(int repr, int64_t n, int d, int k, const void *x, const void *scree
                        (repr == SKM_REPR_LVQ4 && d <= TC_LVQ4_MAX_D) ||
                        (repr == SKM_REPR_SQ8 && d <= TC_SQ8_MAX_D);
     if (!dense) return;
-    const bool pk = repr == SKM_REPR_RBQ1 && !screen && rbq1_packed(d, x);
+    const bool pk = !screen && ((repr == SKM_REPR_RBQ1 && rbq1_packed(d, x)) ||
+                                (repr == SKM_REPR_LVQ4 && lvq4_packed(d, x)));
     if (!screen && !pk) {
         const size_t sb = tc_screen_bytes(repr, n, d, x);
         b.screen = cv.take<uint8_t>(sb);
     }
     const size_t kp = (size_t)cdiv(k, BN) * BN;  // per-centroid records padded to whole tiles
     if (repr == SKM_REPR_LVQ4) {
+        if (pk)  // read packed: per-CTA expansion slots (two per job stream)
+            b.pk_scratch = cv.take<uint8_t>((size_t)std::min<int64_t>(PK_MAX_CTAS, cdiv(n, BM)) * TC_NS[MODE_LVQ4] *
+                                            2 * BM * round16(d));
         b.cs = reinterpret_cast<uint16_t *>(cv.take<uint8_t>((size_t)k * round16(d)));
         b.linfo = cv.take<float4>(k);
         b.rpair_bs = cv.take<float4>(kp / 2);
@@ -2230,7 +2290,8 @@ int tc_assign_lvq4(const skm_data *x, const float *C, int k, int32_t *assign, fl
     const int64_t n = x->n;
     const int d = x->d, dp = round16(d);
     const void *screen = x->screen;
-    if (!screen) {
+    // without a caller copy the codes are read packed where their layout allows
+    if (!screen && !lvq4_packed(d, x->x)) {
         SKM_TRY(tc_screen_prep(x, b.screen, st));
         screen = b.screen;
     }
@@ -2247,8 +2308,14 @@ int tc_assign_lvq4(const skm_data *x, const float *C, int k, int32_t *assign, fl
     p.rinfoq = b.rpair_qn;
     p.lvq = reinterpret_cast<const float4 *>(x->lvq);
     p.d = d;
+    if (v.packed) {
+        p.pk_codes = static_cast<const uint32_t *>(x->x);
+        p.pk_scratch = b.pk_scratch;
+        p.pk_words = lvq4_words(d);
+        p.pk_dp = dp;
+    }
     SKM_TRY(seg_setup(seg, n, p, st));
-    SKM_TRY(launch_tc<MODE_LVQ4>(v.xs, n, dp, d, b.cs, k, p, st));
+    SKM_TRY(launch_tc<MODE_LVQ4>(v.xs, n, dp, d, b.cs, k, p, st, v.packed));
     add_stats_kernel<<<1, 1, 0, st>>>(b.counters, b.stats);
     SKM_CUDA_TRY(launched());
     return SKM_OK;

@@ -224,7 +224,7 @@ static void plan_fit(const skm_data *x, int k, Carver &cv, FitBufs &b) {
     skm_data xs = *x;
     if (x->repr == SKM_REPR_F32 || x->repr == SKM_REPR_BF16) xs.flags |= SKM_FLAG_WARM;  // as skm_fit
     // 1-bit codes the tensor-core kernel reads packed: no copy of the points
-    const bool packed = x->repr == SKM_REPR_RBQ1 && tc_rbq1_reads_packed(x->d, x->x);
+    const bool packed = tc_reads_packed(x->repr, x->d, x->x);
     if (!x->screen && !packed) {
         const size_t sb = tc_screen_bytes(x->repr, x->n, x->d, x->x);
         if (sb) {

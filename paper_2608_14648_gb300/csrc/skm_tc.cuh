@@ -55,9 +55,9 @@ struct TcSeg {
 
 size_t tc_screen_bytes(int repr, int64_t n, int d, const void *x);
 int tc_screen_prep(const skm_data *x, void *screen, cudaStream_t st);
-// whether the 1-bit tensor-core assignment reads these codes packed when
-// no screening copy is given
-bool tc_rbq1_reads_packed(int d, const void *x);
+// whether the 1-bit / LVQ4 tensor-core assignment reads these codes packed
+// when no screening copy is given
+bool tc_reads_packed(int repr, int d, const void *x);
 void tc_plan(int repr, int64_t n, int d, int k, const void *x, const void *screen, bool warm, Carver &cv,
              TcAssignBufs &b);
 int tc_init_stats(TcAssignBufs &b, cudaStream_t st);

@@ -284,3 +284,20 @@ def test_rbq1_packed_reading_needs_no_screen_workspace(skm):
         assert packed < n * d // 4 and copied >= n * d
     # 3 words a row: the copy
     assert L.skm_workspace_size(0, ctypes.byref(data(96, 0x1000, n)), 1000) >= n * 96
+
+
+def test_lvq4_packed_reading_needs_no_screen_workspace(skm):
+    """LVQ4 nibble rows of a multiple of 16 bytes at a 16-byte aligned address
+    are read packed when no e4m3 copy is given (per-CTA expansion slots in
+    the workspace instead of a copy of all points)."""
+    L = skm.lib()
+
+    def data(d, ptr, n):
+        return skm.Data(4, d, n, ptr, None, None, None, None, 0, 0, None, FAKE)
+
+    n = 1_000_000
+    for d in (768, 1024, 992):
+        packed = L.skm_workspace_size(0, ctypes.byref(data(d, 0x1000, n)), 1000)
+        copied = L.skm_workspace_size(0, ctypes.byref(data(d, 0x1004, n)), 1000)
+        assert packed < n * d // 4 and copied >= n * d
+    assert L.skm_workspace_size(0, ctypes.byref(data(1000, 0x1000, n)), 1000) >= n * 1000  # 125 words

@@ -980,7 +980,7 @@ def test_encode_lvq4_half_integer_quotients(skm, d):
 
 
 @pytest.mark.parametrize("n,d,k", [(3000, 768, 300), (777, 33, 7), (500, 64, 1), (1000, 1024, 65),
-                                   (600, 1500, 40), (300, 5, 300), (2100, 128, 513)])
+                                   (600, 1500, 40), (300, 5, 300), (2100, 128, 513), (1300, 992, 300)])
 def test_assign_update_lvq4_bitexact(skm, n, d, k):
     X = _points(n, d, seed=n + 4)
     q = skm.skm_quantize(skm.REPR_LVQ4, X.to(DEV))
@@ -996,6 +996,35 @@ def test_assign_update_lvq4_bitexact(skm, n, d, k):
     Co, co = oracle.lvq4_update(h["codes"], h["fac"], pts.rbq1_exp, ao, C.numpy())
     np.testing.assert_array_equal(counts.cpu().numpy(), co)
     np.testing.assert_array_equal(Cn.cpu().numpy(), Co)
+
+
+@pytest.mark.parametrize("d", [128, 768, 992])
+def test_assign_lvq4_packed_codes_equal_expanded_copy(skm, d):
+    """Without a screening copy the tensor-core kernel reads 16-byte aligned
+    LVQ4 nibble words packed (converter warps expand each point tile through
+    a byte -> two e4m3 codes table); misaligned words or a caller-built copy
+    are read from the e4m3 copy.  All give the oracle's result bit for bit."""
+    n, k = 3001, 260
+    X = _points(n, d, seed=d + 37)
+    q = skm.skm_quantize(skm.REPR_LVQ4, X.to(DEV))
+    pts = skm.lvq4_points(q, d)
+    words = q["codes"].view(torch.int32).reshape(n, -1)
+    W = words.shape[1]
+    buf = torch.zeros(n * W + 1, dtype=torch.int32, device=DEV)
+    buf[1:] = words.reshape(-1)
+    off = buf[1:].view(n, W)  # 4 bytes past a 16-byte boundary
+    assert off.data_ptr() % 16 == 4 and pts.x.data_ptr() % 16 == 0
+    pts_off = skm.Points(skm.REPR_LVQ4, off, d, rbq1_exp=pts.rbq1_exp, lvq=pts.lvq)
+    C = X[synth.forgy_indices(n, k, seed=3)].clone().to(DEV)
+    a, dist = skm.skm_assign(pts, C)
+    a2, dist2 = skm.skm_assign(pts_off, C)
+    a3, dist3 = skm.skm_assign(pts.with_screen(), C)
+    h = _lvq4_host(q, d)
+    ao, do = oracle.lvq4_assign(h["codes"], h["fac"], oracle.lvq4_encode(C.cpu().numpy()))
+    np.testing.assert_array_equal(a.cpu().numpy(), ao)
+    np.testing.assert_array_equal(dist.cpu().numpy(), do)
+    assert torch.equal(a, a2) and torch.equal(dist, dist2)
+    assert torch.equal(a, a3) and torch.equal(dist, dist3)
 
 
 @pytest.mark.parametrize("d", [1024, 777])
