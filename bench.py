@@ -699,8 +699,20 @@ def run_case(args):
         Xb = X.to(torch.bfloat16).view(torch.int16).contiguous()
         pts = skm.Points(skm.REPR_BF16, Xb, d).with_screen()
         C = (Xb[synth.forgy_indices(n, k, seed=0).cuda()].to(torch.int32) << 16).view(torch.float32).contiguous()
-    elif args.case == "assign_prune":  # bf16 points, exact prefix-block pruning
-        Xb = X.to(torch.bfloat16).view(torch.int16).contiguous()
+    elif args.case in ("assign_prune", "assign_prune_front"):  # bf16 points, exact prefix-block pruning
+        if args.case == "assign_prune_front":
+            # the 10M PCA-256 recipe at n points and k = n_comp centroids: 1024
+            # dimensions projected to d with the sample's own PCA, in bf16
+            import dataclasses
+
+            spec = dataclasses.replace(synth.WORKLOADS[HEAD], n=n, k=k, n_comp=k)
+            del X
+            X = synth.workload_points(spec, seed=0, device="cuda")
+            mean, P, _ = skm.skm_pca_fit(X, d)
+            X = skm.skm_project(X, P, mean, out_dtype=skm.DTYPE_BF16).view(torch.int16).contiguous()
+            Xb = X
+        else:
+            Xb = X.to(torch.bfloat16).view(torch.int16).contiguous()
         pts = skm.Points(skm.REPR_BF16, Xb, d, flags=skm.FLAG_PRUNE)
         C = (Xb[synth.forgy_indices(n, k, seed=0).cuda()].to(torch.int32) << 16).view(torch.float32).contiguous()
     else:
@@ -719,6 +731,16 @@ def run_case(args):
         tp[0].record()
         skm.skm_assign(pts.with_flags(0), C, k, want_dist=False)
         tp[1].record()
+    if args.case == "assign_prune_front":
+        # a later Lloyd iteration: centroids after three dense steps, the bound
+        # seeded with the dense assignment (the tensor-core front runs)
+        dense = pts.with_flags(0).with_screen()
+        C, _, _, _, _ = skm.skm_fit(dense, k, 3, C_init=C, want_objective=False, want_dist=False)
+        prev, _ = skm.skm_assign(dense, C, k, want_dist=False)
+        tp = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        tp[0].record()
+        skm.skm_assign(dense, C, k, want_dist=False)
+        tp[1].record()
     skm.skm_assign(pts, C, k, prev_assign=prev, want_dist=False, ws=wsA, out=a)
     torch.cuda.synchronize()
     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
@@ -734,12 +756,15 @@ def run_case(args):
     torch.cuda.synchronize()
     out = {"case": args.case, "n": n, "d": d, "k": k, "reps": args.reps,
            "ms_per_call": e0.elapsed_time(e1) / args.reps}
-    if args.case in ("assign_prune", "assign_prune_sq8"):  # the work the bounds left (last timed call)
+    if args.case in ("assign_prune", "assign_prune_sq8", "assign_prune_front"):  # the work the bounds left
         st = skm.skm_assign_prune_stats(wsA)
         pairs = float(n) * k
         out["first_block_survivors"] = st["prune_first_block"] / pairs
         out["complete_survivors"] = st["prune_complete"] / pairs
         out["later_blocks_per_pair"] = st["prune_blocks"] / pairs
+        if args.case == "assign_prune_front":
+            out["prune_stats"] = st
+            out["dense_screen_ms"] = tp[0].elapsed_time(tp[1])
     if args.case == "assign_f32":  # how often the screen alone decides a row
         _, _, _, _, stats = skm.skm_fit(pts, k, 0, C_init=C, want_objective=False, want_dist=False)
         out["screen_stats"] = stats

@@ -148,7 +148,9 @@ typedef struct skm_stats {
     int64_t fallback_rows;    /* F32/BF16: rows rescanned over all k in fp32  */
     int64_t empty_clusters;   /* after the last update                         */
     int64_t prune_first_block;/* SKM_FLAG_PRUNE: (row, centroid) pairs alive
-                                 after the first 32-dimension block             */
+                                 after the first 32-dimension block (after the
+                                 prune_front_dims dimensions when the
+                                 tensor-core front ran)                        */
     int64_t prune_complete;   /* ... alive after the last block                 */
     double cluster_size_std;  /* population standard deviation of the k
                                  cluster sizes of the final assignment (the
@@ -161,7 +163,18 @@ typedef struct skm_stats {
                                  block partial sums evaluated after the first
                                  block (the executed work beyond the n k first
                                  blocks); 0 for RBQ1, whose checkpoints are
-                                 counted by the two fields above               */
+                                 counted by the two fields above.  With the
+                                 tensor-core front: every block partial sum
+                                 evaluated on CUDA cores (the front's work is
+                                 n k prune_front_dims products)               */
+    int64_t prune_front_dims; /* BF16 with SKM_FLAG_PRUNE and a seed
+                                 assignment: dimensions screened on tensor
+                                 cores for every pair (0: none)                */
+    int64_t prune_rows_finished; /* ... rows whose 2 or more survivors were
+                                 finished on CUDA cores (the rest were decided
+                                 by the front, or:)                            */
+    int64_t prune_rows_full;  /* ... rows pruned over all k on CUDA cores
+                                 (more survivors than the front keeps)         */
 } skm_stats;
 
 const char *skm_last_error(void);
@@ -439,6 +452,16 @@ int skm_screen_prep(const skm_data *x, void *screen, size_t screen_bytes, void *
  *  pruning bound with the distance to its previous centroid (entries outside
  *  [0, k) seed with centroid 0; results do not depend on it).  May alias
  *  `assign`.
+ *  BF16 with SKM_FLAG_PRUNE, prev_assign given, 256 <= d <= 1024, d % 8 == 0
+ *  and x 16-byte aligned: the first 128 dimensions of every pair are screened
+ *  on tensor cores (Section 3.1 "SuperKMeans": a GEMM over the front
+ *  dimensions).  A rigorous lower bound of each pair's pruned distance from
+ *  the bf16 product drops the pairs that cannot beat the seed's distance; a
+ *  row whose one survivor is its seed is decided there, rows with 2..128
+ *  survivors finish on CUDA cores with the same block sums, rows with more
+ *  are pruned over all k.  The result is the same as without the front, bit
+ *  for bit (assignments and distances); the workspace then holds about
+ *  280 bytes per point (the survivor lists).
  * ------------------------------------------------------------------------ */
 int skm_assign(const skm_data *x, const void *C, int k, const int32_t *prev_assign,
                int32_t *assign, float *dist, void *ws, size_t ws_bytes, void *stream);

@@ -80,7 +80,9 @@ class Stats(ctypes.Structure):
     _fields_ = [("rescored_rows", ctypes.c_int64), ("fallback_rows", ctypes.c_int64),
                 ("empty_clusters", ctypes.c_int64), ("prune_first_block", ctypes.c_int64),
                 ("prune_complete", ctypes.c_int64), ("cluster_size_std", ctypes.c_double),
-                ("empty_per_iter", ctypes.c_void_p), ("prune_blocks", ctypes.c_int64)]
+                ("empty_per_iter", ctypes.c_void_p), ("prune_blocks", ctypes.c_int64),
+                ("prune_front_dims", ctypes.c_int64), ("prune_rows_finished", ctypes.c_int64),
+                ("prune_rows_full", ctypes.c_int64)]
 
 
 class HierConfig(ctypes.Structure):
@@ -425,7 +427,8 @@ def skm_assign_prune_stats(ws, stream=None):
     st = Stats()
     _check(lib().skm_assign_prune_stats(_ptr(ws), ws.numel(), ctypes.byref(st), _stream(stream)))
     return {"prune_first_block": st.prune_first_block, "prune_complete": st.prune_complete,
-            "prune_blocks": st.prune_blocks}
+            "prune_blocks": st.prune_blocks, "prune_front_dims": st.prune_front_dims,
+            "prune_rows_finished": st.prune_rows_finished, "prune_rows_full": st.prune_rows_full}
 
 
 def skm_assign_rbq1_noalloc(pts: Points, C, out, dist_out=None, stream=None):
@@ -513,7 +516,8 @@ def skm_fit(pts: Points, k, iters, C_init=None, init_idx=None, want_objective=Tr
     stats = {"rescored_rows": st.rescored_rows, "fallback_rows": st.fallback_rows,
              "empty_clusters": st.empty_clusters, "prune_first_block": st.prune_first_block,
              "prune_complete": st.prune_complete, "prune_blocks": st.prune_blocks,
-             "cluster_size_std": st.cluster_size_std,
+             "prune_front_dims": st.prune_front_dims, "prune_rows_finished": st.prune_rows_finished,
+             "prune_rows_full": st.prune_rows_full, "cluster_size_std": st.cluster_size_std,
              "empty_per_iter": list(empties)[:min(iters, 4096)]}
     return C, assign, dist, (list(obj) if obj is not None else None), stats
 

@@ -62,6 +62,92 @@ __device__ __forceinline__ float block_partial(const float *sx, const float *c, 
     return s;
 }
 
+// One warp prunes the centroid batches [c0, c0 + PR_BATCH) for c0 = c_first,
+// c_first + c_step, ... below k against its running bound (beta, best): per
+// batch, lane l takes the first block of centroids c0 + 32 s + l, the
+// survivors (partial <= beta * slack) are compacted into the warp's queue
+// with __ballot_sync / __popc, each further block re-filters the queue the
+// same way, and the complete candidates' full distances update the bound
+// (ties to the lowest index).  qid / qps: the warp's two queues.
+__device__ __forceinline__ void prune_batches(const float *sx, const float *__restrict__ C, int d, int k, int c_first,
+                                              int c_step, float slack, float &beta, int &best,
+                                              int (&qid)[2][PR_BATCH], float (&qps)[2][PR_BATCH],
+                                              unsigned long long &first_alive, unsigned long long &complete,
+                                              unsigned long long &later) {
+    const int lane = threadIdx.x & 31;
+    const unsigned lt = (1u << lane) - 1u;
+    const int nb = (d + 31) >> 5;
+    for (int c0 = c_first; c0 < k; c0 += c_step) {
+        __syncwarp();  // queue 0 may still be read by the previous batch
+        // first block over the whole batch, survivors compacted into queue 0
+        int cnt = 0;
+        for (int s = 0; s < PR_BATCH / 32; ++s) {
+            const int j = c0 + 32 * s + lane;
+            const float p = (j < k) ? block_partial(sx, C + (int64_t)j * d, d, 0) : INFINITY;
+            const bool alive = p <= beta * slack;
+            const unsigned m = __ballot_sync(0xffffffffu, alive);
+            if (alive) {
+                const int pos = cnt + __popc(m & lt);
+                qid[0][pos] = j;
+                qps[0][pos] = p;
+            }
+            cnt += __popc(m);
+        }
+        first_alive += cnt;
+        int src = 0;
+        for (int b = 1; b < nb && cnt > 0; ++b) {
+            __syncwarp();
+            later += cnt;
+            int ncnt = 0;
+            for (int t0 = 0; t0 < cnt; t0 += 32) {
+                const int t = t0 + lane;
+                const bool valid = t < cnt;
+                const int j = valid ? qid[src][t] : 0;
+                const float p = valid ? qps[src][t] + block_partial(sx, C + (int64_t)j * d, d, b) : INFINITY;
+                const bool alive = valid && p <= beta * slack;
+                const unsigned m = __ballot_sync(0xffffffffu, alive);
+                if (alive) {
+                    const int pos = ncnt + __popc(m & lt);
+                    qid[src ^ 1][pos] = j;
+                    qps[src ^ 1][pos] = p;
+                }
+                ncnt += __popc(m);
+            }
+            cnt = ncnt;
+            src ^= 1;
+        }
+        __syncwarp();
+        complete += cnt;
+        // complete candidates: full distances; keep the smallest (lowest index on ties)
+        for (int t0 = 0; t0 < cnt; t0 += 32) {
+            const int t = t0 + lane;
+            float p = INFINITY;
+            int j = 0x7fffffff;
+            if (t < cnt) {
+                p = qps[src][t];
+                j = qid[src][t];
+            }
+#pragma unroll
+            for (int o = 16; o > 0; o >>= 1) {
+                const float op = __shfl_xor_sync(0xffffffffu, p, o);
+                const int oj = __shfl_xor_sync(0xffffffffu, j, o);
+                if (op < p || (op == p && oj < j)) {
+                    p = op;
+                    j = oj;
+                }
+            }
+            if (p < beta || (p == beta && j < best)) {
+                beta = p;
+                best = j;
+            }
+        }
+    }
+}
+
+// relative rounding of a d-term fp32 sum of non-negative terms is below
+// d * 2^-24; keep anything within twice that of beta
+__device__ __forceinline__ float prune_slack(int d) { return 1.0f + 2.0f * (float)(d + 1) * 0x1p-24f; }
+
 template <typename TX>
 __global__ void __launch_bounds__(PR_WARPS * 32) prune_assign_kernel(
     const TX *__restrict__ X, int64_t n, int d, const float *__restrict__ C, int k,
@@ -71,12 +157,9 @@ __global__ void __launch_bounds__(PR_WARPS * 32) prune_assign_kernel(
     __shared__ int qid[PR_WARPS][2][PR_BATCH];
     __shared__ float qps[PR_WARPS][2][PR_BATCH];
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const unsigned lt = (1u << lane) - 1u;
     float *sx = sx_all[warp];
     const int nb = (d + 31) >> 5;
-    // relative rounding of a d-term fp32 sum of non-negative terms is below
-    // d * 2^-24; keep anything within twice that of beta
-    const float slack = 1.0f + 2.0f * (float)(d + 1) * 0x1p-24f;
+    const float slack = prune_slack(d);
     const int64_t nw = (int64_t)gridDim.x * PR_WARPS;
     unsigned long long first_alive = 0, complete = 0, later = 0;
     for (int64_t row = (int64_t)blockIdx.x * PR_WARPS + warp; row < n; row += nw) {
@@ -87,78 +170,67 @@ __global__ void __launch_bounds__(PR_WARPS * 32) prune_assign_kernel(
         if (best < 0 || best >= k) best = 0;
         float beta = 0.0f;
         for (int b = 0; b < nb; ++b) beta += block_partial(sx, C + (int64_t)best * d, d, b);
-        for (int c0 = 0; c0 < k; c0 += PR_BATCH) {
-            __syncwarp();  // queue 0 may still be read by the previous batch
-            // first block over the whole batch, survivors compacted into queue 0
-            int cnt = 0;
-            for (int s = 0; s < PR_BATCH / 32; ++s) {
-                const int j = c0 + 32 * s + lane;
-                const float p = (j < k) ? block_partial(sx, C + (int64_t)j * d, d, 0) : INFINITY;
-                const bool alive = p <= beta * slack;
-                const unsigned m = __ballot_sync(0xffffffffu, alive);
-                if (alive) {
-                    const int pos = cnt + __popc(m & lt);
-                    qid[warp][0][pos] = j;
-                    qps[warp][0][pos] = p;
-                }
-                cnt += __popc(m);
-            }
-            first_alive += cnt;
-            int src = 0;
-            for (int b = 1; b < nb && cnt > 0; ++b) {
-                __syncwarp();
-                later += cnt;
-                int ncnt = 0;
-                for (int t0 = 0; t0 < cnt; t0 += 32) {
-                    const int t = t0 + lane;
-                    const bool valid = t < cnt;
-                    const int j = valid ? qid[warp][src][t] : 0;
-                    const float p =
-                        valid ? qps[warp][src][t] + block_partial(sx, C + (int64_t)j * d, d, b) : INFINITY;
-                    const bool alive = valid && p <= beta * slack;
-                    const unsigned m = __ballot_sync(0xffffffffu, alive);
-                    if (alive) {
-                        const int pos = ncnt + __popc(m & lt);
-                        qid[warp][src ^ 1][pos] = j;
-                        qps[warp][src ^ 1][pos] = p;
-                    }
-                    ncnt += __popc(m);
-                }
-                cnt = ncnt;
-                src ^= 1;
-            }
-            __syncwarp();
-            complete += cnt;
-            // complete candidates: full distances; keep the smallest (lowest index on ties)
-            for (int t0 = 0; t0 < cnt; t0 += 32) {
-                const int t = t0 + lane;
-                float p = INFINITY;
-                int j = 0x7fffffff;
-                if (t < cnt) {
-                    p = qps[warp][src][t];
-                    j = qid[warp][src][t];
-                }
-#pragma unroll
-                for (int o = 16; o > 0; o >>= 1) {
-                    const float op = __shfl_xor_sync(0xffffffffu, p, o);
-                    const int oj = __shfl_xor_sync(0xffffffffu, j, o);
-                    if (op < p || (op == p && oj < j)) {
-                        p = op;
-                        j = oj;
-                    }
-                }
-                if (p < beta || (p == beta && j < best)) {
-                    beta = p;
-                    best = j;
-                }
-            }
-        }
+        prune_batches(sx, C, d, k, 0, PR_BATCH, slack, beta, best, qid[warp], qps[warp], first_alive, complete,
+                      later);
         if (lane == 0) {
             assign[row] = best;
             if (dist) dist[row] = beta;
         }
     }
     if (counters && lane == 0) {
+        atomicAdd(&counters[0], first_alive);
+        atomicAdd(&counters[1], complete);
+        atomicAdd(&counters[2], later);
+    }
+}
+
+// The same pruning for a list of rows (those the tensor-core front could
+// not keep the survivors of), one CTA of PRC_WARPS warps per row: the warps
+// split the centroid batches, each starting from the row's seed distance
+// beta0 (already computed, the same value as above) and its seed, and the
+// CTA keeps the smallest (distance, index) of the warps' results.
+constexpr int PRC_WARPS = 8;
+__global__ void __launch_bounds__(PRC_WARPS * 32) prune_rows_cta_kernel(
+    const uint16_t *__restrict__ X, int d, const float *__restrict__ C, int k, const int32_t *__restrict__ prev,
+    const float2 *__restrict__ thr, const int32_t *__restrict__ rows, const unsigned long long *__restrict__ nrows,
+    int32_t *__restrict__ assign, float *__restrict__ dist, unsigned long long *__restrict__ counters) {
+    __shared__ float sx[PR_MAX_D];
+    __shared__ int qid[PRC_WARPS][2][PR_BATCH];
+    __shared__ float qps[PRC_WARPS][2][PR_BATCH];
+    __shared__ float wp[PRC_WARPS];
+    __shared__ int wj[PRC_WARPS];
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const float slack = prune_slack(d);
+    const int64_t nr = (int64_t)*nrows;
+    unsigned long long first_alive = 0, complete = 0, later = 0;
+    for (int64_t ri = blockIdx.x; ri < nr; ri += gridDim.x) {
+        const int64_t row = rows[ri];
+        __syncthreads();  // the previous row's sx and results are read
+        for (int i = threadIdx.x; i < d; i += blockDim.x) sx[i] = ldx<uint16_t>(X + row * d + i);
+        __syncthreads();
+        int best = prev ? prev[row] : 0;
+        if (best < 0 || best >= k) best = 0;
+        float beta = thr[row].y;
+        prune_batches(sx, C, d, k, warp * PR_BATCH, PRC_WARPS * PR_BATCH, slack, beta, best, qid[warp], qps[warp],
+                      first_alive, complete, later);
+        if (lane == 0) {
+            wp[warp] = beta;
+            wj[warp] = best;
+        }
+        __syncthreads();
+        if (threadIdx.x == 0) {
+            float bp = wp[0];
+            int bj = wj[0];
+            for (int w = 1; w < PRC_WARPS; ++w)
+                if (wp[w] < bp || (wp[w] == bp && wj[w] < bj)) {
+                    bp = wp[w];
+                    bj = wj[w];
+                }
+            assign[row] = bj;
+            if (dist) dist[row] = bp;
+        }
+    }
+    if (lane == 0 && (first_alive | complete | later)) {
         atomicAdd(&counters[0], first_alive);
         atomicAdd(&counters[1], complete);
         atomicAdd(&counters[2], later);
@@ -470,6 +542,202 @@ __global__ void __launch_bounds__(TP_WARPS * 32) prune_tiled_kernel(
     }
 }
 
+// ------------------------------------------------ tensor-core front (bf16)
+// The seeds' pruned distances and the front's thresholds.  G lanes per row
+// (a power of two at least the number of 32-dimension blocks), lane b
+// computing block b's partial exactly as block_partial does (x_i - c_i then
+// an FMA chain in increasing i), the row's first lane summing the partials
+// in block order: beta0 is the very value the pruning kernels compute for
+// the seed.
+//
+// Threshold: the pruned distance D(x, c) is at least the fp32 partial over
+// the first F dimensions (fp32 sums of non-negative terms never decrease),
+// which is at least (1 - gamma) S_F, S_F = sum_{i < F} (x_i - c_i)^2 =
+// ||x_F||^2 + s_F with s_F = ||c_F||^2 - 2 <x_F, c_F>, gamma = (34 + F/32)
+// 2^-24 (one rounding per subtraction and square, 32 per block chain, one
+// per block sum).  The tensor-core front evaluates s~_F with |s~_F - s_F| <=
+// 2 ||x_F|| h'_j + z_j <= W = 2 ||x_F|| max h' + max z (the screen's interval
+// with prefix norms; bf16 points are their own operand).  A centroid with
+// s~_F > thr = beta0 slack (1 + 2^-16) - ||x_F||^2 + W (each step rounded
+// outwards; 2^-16 covers 1 / (1 - gamma) and the rounding of beta0 slack)
+// therefore has D(x, c) > fl(beta0 slack) >= the row's minimum and is
+// dropped: the pruning kernels, seeded alike, never complete it either
+// (slack is theirs).  A non-finite seed distance keeps everything (the row then
+// overflows to the full pruning).
+// One 32-dimension block of (x_i - c_i)^2 for a lane: x from bf16 (16-byte
+// loads), c from fp32 (16-byte loads), every load issued before the chain;
+// the sum runs in increasing i as in block_partial.  q (when wanted) gets the
+// sum of x_i^2 over the block.  m = dimensions in the block (32 unless it is
+// the ragged last one).
+__device__ __forceinline__ float block_bf16(const uint16_t *xr, const float *cr, int m, bool want_q, float &q) {
+    float part = 0.0f;
+    q = 0.0f;
+    if (m == 32) {
+        uint4 xw[4];
+        float4 cv[8];
+#pragma unroll
+        for (int u = 0; u < 4; ++u) xw[u] = __ldg(reinterpret_cast<const uint4 *>(xr) + u);
+#pragma unroll
+        for (int u = 0; u < 8; ++u) cv[u] = __ldg(reinterpret_cast<const float4 *>(cr) + u);
+#pragma unroll
+        for (int u = 0; u < 8; ++u) {
+            const uint32_t w0 = (u & 1) ? xw[u >> 1].z : xw[u >> 1].x;
+            const uint32_t w1 = (u & 1) ? xw[u >> 1].w : xw[u >> 1].y;
+            const float xs[4] = {__uint_as_float(w0 << 16), __uint_as_float(w0 & 0xffff0000u),
+                                 __uint_as_float(w1 << 16), __uint_as_float(w1 & 0xffff0000u)};
+            const float cs[4] = {cv[u].x, cv[u].y, cv[u].z, cv[u].w};
+#pragma unroll
+            for (int h = 0; h < 4; ++h) {
+                const float t = __fsub_rn(xs[h], cs[h]);
+                part = __fmaf_rn(t, t, part);
+                if (want_q) q = __fmaf_rn(xs[h], xs[h], q);
+            }
+        }
+    } else {
+        for (int i = 0; i < m; ++i) {
+            const float xv = __uint_as_float(((uint32_t)__ldg(xr + i)) << 16);
+            const float t = __fsub_rn(xv, __ldg(cr + i));
+            part = __fmaf_rn(t, t, part);
+            if (want_q) q = __fmaf_rn(xv, xv, q);
+        }
+    }
+    return part;
+}
+
+__global__ void front_prep_kernel(const uint16_t *__restrict__ X, int64_t n, int d, int F, int G,
+                                  const float *__restrict__ C, int k, const int32_t *__restrict__ prev,
+                                  const float *__restrict__ hz, float2 *__restrict__ thr,
+                                  unsigned long long *__restrict__ ctr) {
+    const int lane = threadIdx.x & 31;
+    const int sub = lane / G, b = lane % G;
+    const int rpw = 32 / G;  // rows per warp
+    const int nb = (d + 31) >> 5;
+    const int64_t warp = (blockIdx.x * (int64_t)blockDim.x + threadIdx.x) >> 5;
+    const int64_t nw = ((int64_t)gridDim.x * blockDim.x) >> 5;
+    if (blockIdx.x == 0 && threadIdx.x == 0) {
+        ctr[3] = (unsigned long long)F;
+        ctr[9] = (unsigned long long)k;
+    }
+    const float H = __ldg(hz), Z = __ldg(hz + 1);
+    const float slack = prune_slack(d);
+    const float K1 = __fmul_ru(slack, 1.0f + 0x1p-16f);
+    for (int64_t r0 = warp * rpw; r0 < n; r0 += nw * rpw) {
+        const int64_t row = r0 + sub;
+        const bool act = row < n;
+        int seed = act && prev ? __ldg(prev + row) : 0;
+        if (seed < 0 || seed >= k) seed = 0;
+        float part = 0.0f, q = 0.0f;
+        if (act && b < nb)
+            part = block_bf16(X + row * d + 32 * b, C + (int64_t)seed * d + 32 * b, min(32, d - 32 * b), 32 * b < F,
+                              q);
+        // the row's blocks in order (every lane of the group forms the same sum)
+        float beta0 = __shfl_sync(0xffffffffu, part, 0, G);
+        for (int t = 1; t < nb; ++t) beta0 = __fadd_rn(beta0, __shfl_sync(0xffffffffu, part, t, G));
+        for (int o = G >> 1; o > 0; o >>= 1) q = __fadd_rn(q, __shfl_xor_sync(0xffffffffu, q, o, G));
+        if (act && b == 0) {
+            // q: fp32 sum of F exact squares, relative error far below (F + 8) 2^-23
+            const float grow = (float)(F + 8) * 0x1p-23f;
+            const float xn_up = __fsqrt_ru(__fmul_ru(q, 1.0f + grow));
+            const float xn2_lo = __fmul_rd(q, 1.0f - grow);
+            const float W = __fmaf_ru(2.0f * xn_up, H, Z);
+            float t = __fadd_ru(__fsub_ru(__fmul_ru(beta0, K1), xn2_lo), W);
+            t = __fadd_ru(t, 0x1p-100f);
+            if (!(t == t) || !(beta0 < INFINITY)) t = INFINITY;
+            thr[row] = make_float2(t, beta0);
+        }
+    }
+}
+
+// Rows the front left with 2 .. cap survivors: each survivor's pruned
+// distance, G lanes per survivor (lane b: block b, block_bf16 as in the
+// seed pass, the group summing the partials in block order: the very value
+// of the pruning kernels), 32 / G survivors a round; the smallest (lowest
+// index on ties) is the row's argmin, the seed (on the list, at exactly
+// beta0) guaranteeing one.  A survivor is complete when its distance is
+// within the seed distance times the slack (its partial sums never exceed
+// the full one).  One warp per row.
+__global__ void __launch_bounds__(256) prune_finish_kernel(
+    const uint16_t *__restrict__ X, int d, int G, const float *__restrict__ C, const float2 *__restrict__ thr,
+    const uint16_t *__restrict__ cand, const int32_t *__restrict__ cnt, int cap, int nsub,
+    const int32_t *__restrict__ perm, const int32_t *__restrict__ rows, const unsigned long long *__restrict__ nrows,
+    int32_t *__restrict__ assign, float *__restrict__ dist, unsigned long long *__restrict__ ctr) {
+    const int lane = threadIdx.x & 31;
+    const int slot = lane / G, b = lane % G, S = 32 / G;
+    const int nb = (d + 31) >> 5;
+    const float slack = prune_slack(d);
+    const int64_t nr = (int64_t)*nrows;
+    const int64_t warp = (blockIdx.x * (int64_t)blockDim.x + threadIdx.x) >> 5;
+    const int64_t nw = ((int64_t)gridDim.x * blockDim.x) >> 5;
+    unsigned long long complete = 0, blocks = 0;
+    for (int64_t ri = warp; ri < nr; ri += nw) {
+        const int64_t row = __ldg(rows + ri);
+        const float lim = __ldg(&thr[row].y) * slack;
+        const uint32_t pc = (uint32_t)__ldg(cnt + row);
+        const int csub = cap / nsub;
+        const int c0 = min((int)(pc & 255u), csub);
+        const int c1 = nsub > 1 ? min((int)((pc >> 8) & 255u), csub) : 0;
+        const int c2 = nsub > 2 ? min((int)((pc >> 16) & 255u), csub) : 0;
+        const int c3 = nsub > 3 ? min((int)(pc >> 24), csub) : 0;
+        const int tot = c0 + c1 + c2 + c3;
+        float bp = INFINITY;
+        int bj = 0x7fffffff;
+        for (int t0 = 0; t0 < tot; t0 += S) {
+            int t = t0 + slot, h = 0;
+            const bool valid = t < tot;
+            if (t >= c0) {  // sub-list h and the position in it
+                t -= c0;
+                h = 1;
+                if (t >= c1) {
+                    t -= c1;
+                    h = 2;
+                    if (t >= c2) {
+                        t -= c2;
+                        h = 3;
+                    }
+                }
+            }
+            const int j = valid ? __ldg(perm + __ldg(cand + row * cap + h * csub + t)) : 0;
+            float part = 0.0f, q;
+            if (valid && b < nb)
+                part = block_bf16(X + row * d + 32 * b, C + (int64_t)j * d + 32 * b, min(32, d - 32 * b), false, q);
+            float D = __shfl_sync(0xffffffffu, part, 0, G);
+            for (int u = 1; u < nb; ++u) D = __fadd_rn(D, __shfl_sync(0xffffffffu, part, u, G));
+            if (valid && b == 0) {
+                blocks += (unsigned long long)nb;
+                if (D <= lim) {
+                    ++complete;
+                    if (D < bp || (D == bp && j < bj)) {
+                        bp = D;
+                        bj = j;
+                    }
+                }
+            }
+        }
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) {
+            const float op = __shfl_xor_sync(0xffffffffu, bp, o);
+            const int oj = __shfl_xor_sync(0xffffffffu, bj, o);
+            if (op < bp || (op == bp && oj < bj)) {
+                bp = op;
+                bj = oj;
+            }
+        }
+        if (lane == 0) {
+            assign[row] = bj;
+            if (dist) dist[row] = bp;
+        }
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+        complete += __shfl_xor_sync(0xffffffffu, complete, o);
+        blocks += __shfl_xor_sync(0xffffffffu, blocks, o);
+    }
+    if (lane == 0 && (complete | blocks)) {
+        atomicAdd(&ctr[1], complete);
+        atomicAdd(&ctr[2], blocks);
+    }
+}
+
 }  // namespace
 
 cudaError_t launch_prune_assign_sq8(const uint8_t *X, int64_t n, int d, const uint8_t *C, int k, const int32_t *prev,
@@ -512,6 +780,44 @@ cudaError_t launch_prune_assign(const void *X, int x_is_bf16, int64_t n, int d, 
     else
         prune_assign_kernel<float><<<(int)blocks, PR_WARPS * 32, 0, st>>>(
             static_cast<const float *>(X), n, d, C, k, prev, assign, dist, counters);
+    return launched();
+}
+
+cudaError_t launch_prune_rows_cta(const uint16_t *X, int d, const float *C, int k, const int32_t *prev,
+                                  const float2 *thr, const int32_t *rows, const unsigned long long *nrows,
+                                  int32_t *assign, float *dist, unsigned long long *counters, cudaStream_t st) {
+    if (d > PR_MAX_D) return cudaErrorInvalidValue;
+    prune_rows_cta_kernel<<<152 * 4, PRC_WARPS * 32, 0, st>>>(X, d, C, k, prev, thr, rows, nrows, assign, dist,
+                                                              counters);
+    return launched();
+}
+
+cudaError_t launch_prune_front_prep(const uint16_t *X, int64_t n, int d, int F, const float *C, int k,
+                                    const int32_t *prev, const float *hz, float2 *thr, unsigned long long *ctr,
+                                    cudaStream_t st) {
+    const int nb = (d + 31) >> 5;
+    int G = 1;
+    while (G < nb) G <<= 1;
+    if (G > 32 || F % 32 != 0 || F > d || (d % 8) != 0) return cudaErrorInvalidValue;
+    const int64_t per_block = 256 / G;  // rows per block of 256 threads
+    int64_t blocks = (n + per_block - 1) / per_block;
+    if (blocks > 152 * 16) blocks = 152 * 16;
+    if (blocks < 1) blocks = 1;
+    front_prep_kernel<<<(int)blocks, 256, 0, st>>>(X, n, d, F, G, C, k, prev, hz, thr, ctr);
+    return launched();
+}
+
+cudaError_t launch_prune_finish(const uint16_t *X, int d, const float *C, const float2 *thr, const uint16_t *cand,
+                                const int32_t *cnt, int cap, int nsub, const int32_t *perm, const int32_t *rows,
+                                const unsigned long long *nrows, int32_t *assign, float *dist,
+                                unsigned long long *ctr, cudaStream_t st) {
+    const int nb = (d + 31) >> 5;
+    int G = 1;
+    while (G < nb) G <<= 1;
+    if (G > 32 || (d % 8) != 0 || nsub < 1 || nsub > 4 || cap % nsub != 0 || cap / nsub > 255)
+        return cudaErrorInvalidValue;
+    prune_finish_kernel<<<152 * 8, 256, 0, st>>>(X, d, G, C, thr, cand, cnt, cap, nsub, perm, rows, nrows, assign,
+                                                 dist, ctr);
     return launched();
 }
 

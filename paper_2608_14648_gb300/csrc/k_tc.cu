@@ -66,10 +66,10 @@ constexpr int64_t WARM_MAGIC = 0x534b4d5741524d31LL;
 constexpr int TCAND = 4;
 constexpr unsigned long long WAIT_LIMIT_NS = 2000000000ull;  // 2 s per barrier wait
 
-enum { MODE_SCREEN = 0, MODE_SQ8 = 1, MODE_RBQ1 = 2, MODE_LVQ4 = 3, MODE_GEMM = 4 };
+enum { MODE_SCREEN = 0, MODE_SQ8 = 1, MODE_RBQ1 = 2, MODE_LVQ4 = 3, MODE_GEMM = 4, MODE_PFRONT = 5 };
 // Epilogue warps per TMEM lane quarter, by mode.  Every CTA works alone
 // (no thread-block clusters): it loads its own centroid slices.
-constexpr int TC_NH[5] = {4, 4, 4, 4, 4};
+constexpr int TC_NH[6] = {4, 4, 4, 4, 4, 4};
 // Job streams per CTA, by mode.  NS = 2: the CTA's point tiles form two
 // streams whose jobs the MMA warp issues alternately, each into its own TMEM
 // accumulator, each drained by its own half of the epilogue warps; an
@@ -79,7 +79,7 @@ constexpr int TC_NH[5] = {4, 4, 4, 4, 4};
 // records.)  Measured at 1M x 1000 x 768 against one stream: 1-bit 0.508 vs
 // 0.574 ms, LVQ4 0.532 vs 0.575, fp32 screen 0.99 vs 1.02, SQ8 (with NH = 4)
 // 0.847 vs 0.882.
-constexpr int TC_NS[5] = {2, 2, 2, 2, 2};
+constexpr int TC_NS[6] = {2, 2, 2, 2, 2, 2};
 // GEMM mode (the projection Y = (X - mean) P in fp32 accuracy from bf16
 // parts x = x1 + x2 + x3, P = p1 + p2 + p3): K segments of (A part, B part),
 // the smallest products first; parts i + j > 4 (below 2^-24 relative) are left
@@ -97,6 +97,14 @@ constexpr int f8_cw() { return MODE == 3 /* MODE_LVQ4 */ ? 32 : 16; }
 // packed FMA per column pair: 32 is 2-4% faster there (C1 1.014 vs 1.032 ms,
 // C4 38.1 vs 39.7 ms).
 constexpr int SCR_CW = 32;
+// PFRONT: the tensor-core front of exact dimension pruning takes the first
+// PF_DIMS dimensions; each row keeps at most PF_CAP survivors (PF_CAP / NHG
+// per column slice of the epilogue, as 16-bit sorted positions, k <= 65536),
+// more send it to the CUDA-core pruning over all k.  Measured on the 10M x 256 PCA workload (k = 10,000, bound from
+// the previous centroid): 1.3 survivors a row after 128 dimensions (99.9% of
+// rows at most 37), 80 after 64 (1% of rows above 2,000).
+constexpr int PF_DIMS = 128;
+constexpr int PF_CAP = 128;
 // the e4m3 (kind::f8f6f4) modes: 128 elements per 128-byte K slice
 template <int MODE>
 constexpr bool f8_mode() { return MODE == MODE_RBQ1 || MODE == MODE_LVQ4; }
@@ -176,6 +184,22 @@ struct TcParams {
     void *y;
     int y_bf16;
     int ydout;
+    // PFRONT: per row (threshold on s~ over the front dimensions, the seed's
+    // pruned distance), survivor lists [n][PF_CAP] (sorted positions, one
+    // sub-list of PF_CAP / NHG per column slice), per listed row the
+    // sub-lists' counts (8 bits each), the seed centroids (NULL: centroid 0)
+    // and the pruning counters ([0] pairs alive after the front, [4] rows
+    // listed for the CUDA-core finish, [5] rows whose lists overflowed)
+    const float2 *pf_thr;
+    uint16_t *pf_cand;
+    // PFRONT: the centroid operand and records are sorted by ||c_F||^2
+    // (pf_perm: sorted position -> centroid); pf_cmin: per 32-column chunk of
+    // sorted positions, the smallest ||c_F||^2
+    const int32_t *pf_perm;
+    const float *pf_cmin;
+    int32_t *pf_cnt;
+    const int32_t *pf_prev;
+    unsigned long long *pf_ctr;
     // Fault injection (0 = off): the producer first waits this long on a
     // barrier that nothing arrives on, so the launch gives up before it has
     // loaded anything and reports through the abort flag.
@@ -356,6 +380,12 @@ __device__ __forceinline__ float fmin3(float a, float b, float c) {
     return r;
 }
 
+__device__ __forceinline__ float fmax3(float a, float b, float c) {
+    float r;
+    asm("max.f32 %0, %1, %2, %3;" : "=f"(r) : "f"(a), "f"(b), "f"(c));
+    return r;
+}
+
 // v[i] for a lane-dependent i in [0, 32): binary select tree (no local memory).
 __device__ __forceinline__ uint32_t pick32(const uint32_t (&v)[32], int i) {
     uint32_t w16[16], w8[8], w4[4], w2[2];
@@ -480,8 +510,10 @@ __global__ void __launch_bounds__(tc_threads<NH, PK>(), 1)
     tc_assign_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                      const TcParams p) {
     static_assert(NS == 1 || (NS == 2 && NH % 2 == 0), "two job streams: two epilogue groups");
-    static_assert(NS == 1 || MODE == MODE_GEMM || epi_threads<NH>() / NS >= (MODE == MODE_SCREEN ? 128 : 256),
+    static_assert(NS == 1 || MODE == MODE_GEMM ||
+                      epi_threads<NH>() / NS >= (MODE == MODE_SCREEN || MODE == MODE_PFRONT ? 128 : 256),
                   "records staged by one epilogue group");
+    static_assert(MODE != MODE_PFRONT || !SEG, "the pruning front has no segmented variant");
     extern __shared__ uint8_t smem_raw[];
     const uint32_t raw = smem_u32(smem_raw);
     const uint32_t base = (raw + 1023u) & ~1023u;
@@ -524,7 +556,7 @@ __global__ void __launch_bounds__(tc_threads<NH, PK>(), 1)
         }
         for (int b = 0; b < 2; ++b) {
             mbar_init(tfull_bar(b), 1);
-            mbar_init(tempty_bar(b), epi_threads<NH>() / NS);
+            mbar_init(tempty_bar(b), epi_threads<NH>() / NS / 32);  // one arrival per epilogue warp
         }
         mbar_init(drain_bar, 1);
         mbar_init(inject_bar, 1);
@@ -874,10 +906,12 @@ __global__ void __launch_bounds__(tc_threads<NH, PK>(), 1)
         float2 pre2 = make_float2(0.f, 0.f);
         int32_t pre1 = 0;
         auto rec_load = [&](int ctn) {
-            if (MODE == MODE_SCREEN) {
+            if (MODE == MODE_SCREEN || MODE == MODE_PFRONT) {
                 if (te < 128) {
                     const float4 ci = __ldg(p.cinfo + ctn * 128 + te);
                     pre2 = make_float2(ci.x, ci.y);
+                } else if (MODE == MODE_PFRONT && te < 130) {  // the tile's 8 chunk minima
+                    pre4 = __ldg(reinterpret_cast<const float4 *>(p.pf_cmin + ctn * 8) + (te - 128));
                 }
             } else if (f8_mode<MODE>()) {
                 if (te < 128) pre4 = __ldg(p.rinfo + ctn * 128 + te);
@@ -888,8 +922,9 @@ __global__ void __launch_bounds__(tc_threads<NH, PK>(), 1)
         };
         auto rec_store = [&](uint32_t buf) {
             uint8_t *rb = rec_base + buf * REC_BYTES;
-            if (MODE == MODE_SCREEN) {
+            if (MODE == MODE_SCREEN || MODE == MODE_PFRONT) {
                 if (te < 128) reinterpret_cast<float2 *>(rb)[te] = pre2;
+                else if (MODE == MODE_PFRONT && te < 130) reinterpret_cast<float4 *>(rb + 1024)[te - 128] = pre4;
             } else if (f8_mode<MODE>()) {
                 if (te < 256) reinterpret_cast<float4 *>(rb)[te] = pre4;
             } else if (MODE == MODE_SQ8) {
@@ -905,6 +940,7 @@ __global__ void __launch_bounds__(tc_threads<NH, PK>(), 1)
         // in the named barriers, so the other epilogue warps never wait on it.
         bool dead = false;
         uint32_t job = 0;  // jobs of this group so far (NS = 1: of the CTA)
+        unsigned long long pf_alive = 0;  // PFRONT: survivors of this thread's rows
         for (int64_t g = g0 + grp * gstep; g < ngroups; g += NS * gstep) {
             const int64_t rt = g;
             const int64_t row = rt * BM + rin;
@@ -915,6 +951,15 @@ __global__ void __launch_bounds__(tc_threads<NH, PK>(), 1)
             float fbest = INFINITY;
             float a2 = 0.0f, w2 = 0.0f, rnx2 = 0.0f, rf2 = 0.0f, rpc = 0.0f;
             int32_t nxr = 0;
+            // PFRONT: survive iff s~ <= pthr; this slice's sub-list and count
+            constexpr int PF_SUB = PF_CAP / NHG;
+            float pthr = -INFINITY;
+            int pcnt = 0;
+            uint16_t *pf_list = nullptr;
+            if (MODE == MODE_PFRONT && valid) {
+                pthr = p.pf_thr[row].x;
+                pf_list = p.pf_cand + row * PF_CAP + slice * PF_SUB;
+            }
             // segmented mode: this row's centroid range (ids clamped into bounds)
             int cb = 0, ce = 0x7fffffff;
             if (SEG && valid) {
@@ -1123,6 +1168,50 @@ __global__ void __launch_bounds__(tc_threads<NH, PK>(), 1)
                             tmem_wait16(va);
                         }
                     }
+                } else if (MODE == MODE_PFRONT) {
+                    // Columns are centroids sorted by ||c_F||^2.  Per 32-column
+                    // chunk: a = the largest accumulator (three-input maxima), and
+                    // fl(cmin - 2 a) <= fl(||c_j||^2 - 2 acc_j) = s~_j for every
+                    // column (rounding is monotone), so a chunk with fl(cmin - 2 a)
+                    // > pthr has no survivor.  Otherwise (rare) each column's s~ is
+                    // formed and those <= pthr are listed (sorted positions).
+                    // Records past k have ||c_F||^2 = +inf.  The slices take
+                    // alternate chunks (neighbouring positions, which similar
+                    // survivors tend to share, go to different sub-lists).
+                    const float *cmins = reinterpret_cast<const float *>(rbuf + 1024);
+                    const uint32_t tbase = tmem + ((uint32_t)(q * 32) << 16) + b * BN;
+#pragma unroll 1
+                    for (int c = 0; c < SW / 32; ++c) {
+                        const int cc = (NHG * c + slice) * 32;  // column offset within the tile
+                        const int j0 = ct * BN + cc;
+                        if (j0 >= p.k) break;  // warp-uniform
+                        uint32_t v[32];
+                        tmem_ld32(tbase + cc, v);
+                        auto f = [&](int i) { return __uint_as_float(v[i]); };
+                        float m[11];
+#pragma unroll
+                        for (int t = 0; t < 10; ++t) m[t] = fmax3(f(3 * t), f(3 * t + 1), f(3 * t + 2));
+                        m[10] = fmaxf(f(30), f(31));
+                        const float amax = fmax3(fmax3(m[0], m[1], m[2]), fmax3(m[3], m[4], m[5]),
+                                                 fmax3(fmax3(m[6], m[7], m[8]), m[9], m[10]));
+                        if (__fmaf_rn(-2.0f, amax, cmins[cc >> 5]) <= pthr && pf_list) {
+                            uint32_t mask = 0;
+#pragma unroll
+                            for (int i = 0; i < 32; i += 4) {
+                                const float4 c4 = reinterpret_cast<const float4 *>(rbuf)[(cc + i) >> 2];
+                                mask |= (__fmaf_rn(-2.0f, f(i), c4.x) <= pthr ? 1u : 0u) << i;
+                                mask |= (__fmaf_rn(-2.0f, f(i + 1), c4.y) <= pthr ? 2u : 0u) << i;
+                                mask |= (__fmaf_rn(-2.0f, f(i + 2), c4.z) <= pthr ? 4u : 0u) << i;
+                                mask |= (__fmaf_rn(-2.0f, f(i + 3), c4.w) <= pthr ? 8u : 0u) << i;
+                            }
+                            while (mask) {
+                                const int i = __ffs(mask) - 1;
+                                mask &= mask - 1u;
+                                if (pcnt < PF_SUB) pf_list[pcnt] = (uint16_t)(j0 + i);
+                                ++pcnt;
+                            }
+                        }
+                    }
                 } else if (f8_mode<MODE>()) {
                     // e4m3 modes: chunks of F8_CW columns (F8_CW = 16: the next
                     // chunk's TMEM load in flight while this one is evaluated)
@@ -1230,8 +1319,11 @@ __global__ void __launch_bounds__(tc_threads<NH, PK>(), 1)
                         }
                     }
                 }
+                // the warp's TMEM loads are complete (each thread waited on
+                // them); one arrival for the warp releases its share
                 tc_fence_before();
-                mbar_arrive(tempty_bar(b));
+                __syncwarp();
+                if (lane == 0) mbar_arrive(tempty_bar(b));
             }
             // merge the column slices of each row: slices 1.. publish, slice 0 finishes
             // (single buffer: a publisher rewrites its slot only at the end of
@@ -1251,13 +1343,44 @@ __global__ void __launch_bounds__(tc_threads<NH, PK>(), 1)
                 } else if (MODE == MODE_SQ8) {
                     slot[0] = (uint32_t)best;
                     slot[1] = (uint32_t)besti;
+                } else if (MODE == MODE_PFRONT) {
+                    slot[0] = (uint32_t)pcnt;
                 } else {
                     slot[0] = __float_as_uint(fbest);
                     slot[1] = (uint32_t)besti;
                 }
             }
             asm volatile("bar.sync %0, %1;" ::"r"(NS == 2 ? 4 + grp : 1), "n"(GT) : "memory");
-            if (slice == 0 && valid && !dead) {
+            if (MODE == MODE_PFRONT && slice == 0 && valid && !dead) {
+                // The row's survivors: one (the seed, whose pruned distance
+                // every pruned pair provably exceeds) decides the row; 2 ..
+                // PF_CAP go to the CUDA-core finish; more, or none
+                // (impossible while the bounds hold), to pruning over all k.
+                int tot = pcnt, one = pcnt == 1 ? 0 : -1;
+                bool over = pcnt > PF_SUB;
+                uint32_t packed = (uint32_t)min(pcnt, 255);
+#pragma unroll
+                for (int h = 1; h < NHG; ++h) {
+                    const int ch = (int)merge[((h - 1) * BM + rin) * MW];
+                    if (ch == 1) one = h;
+                    tot += ch;
+                    over = over || ch > PF_SUB;
+                    packed |= (uint32_t)min(ch, 255) << (8 * h);
+                }
+                pf_alive += (unsigned long long)tot;
+                int seed = p.pf_prev ? p.pf_prev[row] : 0;
+                seed = (seed < 0 || seed >= p.k) ? 0 : seed;
+                if (!over && tot == 1 && one >= 0 && p.pf_perm[p.pf_cand[row * PF_CAP + one * PF_SUB]] == seed) {
+                    p.assign[row] = seed;
+                    if (p.dist) p.dist[row] = p.pf_thr[row].y;
+                } else if (!over && tot >= 2) {
+                    p.pf_cnt[row] = (int32_t)packed;
+                    p.resc_rows[atomicAdd(p.pf_ctr + 4, 1ull)] = (int32_t)row;
+                } else {
+                    p.fall_rows[atomicAdd(p.pf_ctr + 5, 1ull)] = (int32_t)row;
+                }
+            }
+            if (MODE != MODE_PFRONT && slice == 0 && valid && !dead) {
                 // slices in increasing column order; ties resolve to the lower index
 #pragma unroll
                 for (int h = 1; h < NHG; ++h) {
@@ -1354,6 +1477,11 @@ __global__ void __launch_bounds__(tc_threads<NH, PK>(), 1)
                     if (p.dist) p.dist[row] = fbest;
                 }
             }
+        }
+        if (MODE == MODE_PFRONT) {
+#pragma unroll
+            for (int o = 16; o > 0; o >>= 1) pf_alive += __shfl_xor_sync(0xffffffffu, pf_alive, o);
+            if (lane == 0 && pf_alive) atomicAdd(p.pf_ctr, pf_alive);
         }
     }
     tc_fence_before();
@@ -1474,7 +1602,9 @@ __global__ void screen_prep_sq8_kernel(const uint8_t *__restrict__ X, int64_t n,
 // h' = e + (eps_acc + eps_s) (||c|| + e) + rho_max ||c||, e = ||c~ - c||,
 // z = eps_s ||c||^2, where rho_max >= ||x~ - x|| / ||x~|| over all points, so
 // |s~ - s| <= 2 ||x~|| h' + z = w (the half-width of the pair's interval).
-// Records j in [k, kp) get ||c||^2 = +inf so they never matter.  Layout:
+// Records j in [k, kp) get ||c||^2 = +inf so they never matter.  The operand
+// and the records cover the first dr dimensions (dr = d, or the pruning
+// front's prefix).  Layout:
 // column pair p = (2p, 2p+1) -> cinfo[p] = (||c||^2 x2, h' x2), cinfoz[p] = (z x2);
 // hz_bits (zeroed by the caller) receives max h' and max z over j < k.
 //
@@ -1484,7 +1614,7 @@ __global__ void screen_prep_sq8_kernel(const uint8_t *__restrict__ X, int64_t n,
 // publishes in *warm_ok whether the stamp names this n, d and k (the bounds
 // and cprev then belong to these points) and clears the stamp until this
 // call completes.
-__global__ void cprep_f32_kernel(const float *__restrict__ C, int k, int kp, int d, int dp,
+__global__ void cprep_f32_kernel(const float *__restrict__ C, int k, int kp, int d, int dp, int dr,
                                  float eps_acc, float eps_s, const float *__restrict__ rho_max,
                                  __nv_bfloat16 *__restrict__ cs, float4 *__restrict__ cinfo,
                                  float2 *__restrict__ cinfoz, unsigned int *__restrict__ hz_bits,
@@ -1511,13 +1641,16 @@ __global__ void cprep_f32_kernel(const float *__restrict__ C, int k, int kp, int
             continue;
         }
         double c2 = 0.0, e2 = 0.0, p2 = 0.0, dd = 0.0, dn = 0.0;
-        for (int i = lane; i < d; i += 32) {
+        const int iend = cprev ? d : dr;
+        for (int i = lane; i < iend; i += 32) {
             const float c = C[(int64_t)j * d + i];
-            const __nv_bfloat16 cb = __float2bfloat16_rn(c);
-            cs[(int64_t)j * dp + i] = cb;
-            const double cf = (double)__bfloat162float(cb);
-            c2 += (double)c * (double)c;
-            e2 += (cf - (double)c) * (cf - (double)c);
+            if (i < dr) {
+                const __nv_bfloat16 cb = __float2bfloat16_rn(c);
+                cs[(int64_t)j * dp + i] = cb;
+                const double cf = (double)__bfloat162float(cb);
+                c2 += (double)c * (double)c;
+                e2 += (cf - (double)c) * (cf - (double)c);
+            }
             if (cprev) {
                 const double cq = (double)cprev[(int64_t)j * d + i];
                 p2 += cq * cq;
@@ -1553,6 +1686,123 @@ __global__ void cprep_f32_kernel(const float *__restrict__ C, int k, int kp, int
             // maxima over the centroids (non-negative: bits order like values)
             atomicMax(hz_bits, __float_as_uint(hf));
             atomicMax(hz_bits + 1, __float_as_uint(zf1));
+        }
+    }
+}
+
+// Pruning front: the centroids' positions sorted (by buckets) by ||c_F||^2,
+// so that the 32 columns of a chunk have nearly the same norm.  One block:
+// the finite keys' range, PF_NB equal buckets, an exclusive scan of their
+// counts, then each centroid takes the next position of its bucket (the
+// order within a bucket is whatever the atomics give: the survivors' lists
+// then differ in order only, which the argmin does not see).
+constexpr int PF_NB = 4096;
+__global__ void __launch_bounds__(1024) pf_sort_kernel(const float4 *__restrict__ cinfo, int k,
+                                                       int32_t *__restrict__ perm) {
+    __shared__ unsigned int cnt[PF_NB];
+    __shared__ float red[2][32];
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    const float *cf = reinterpret_cast<const float *>(cinfo);
+    auto key = [&](int j) { return cf[4 * (j >> 1) + (j & 1)]; };
+    float lo = INFINITY, hi = -INFINITY;
+    for (int j = threadIdx.x; j < k; j += blockDim.x) {
+        const float v = key(j);
+        if (v < INFINITY && v == v) {
+            lo = fminf(lo, v);
+            hi = fmaxf(hi, v);
+        }
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+        lo = fminf(lo, __shfl_xor_sync(0xffffffffu, lo, o));
+        hi = fmaxf(hi, __shfl_xor_sync(0xffffffffu, hi, o));
+    }
+    if (lane == 0) {
+        red[0][warp] = lo;
+        red[1][warp] = hi;
+    }
+    for (int b = threadIdx.x; b < PF_NB; b += blockDim.x) cnt[b] = 0u;
+    __syncthreads();
+    lo = red[0][lane];
+    hi = red[1][lane];
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+        lo = fminf(lo, __shfl_xor_sync(0xffffffffu, lo, o));
+        hi = fmaxf(hi, __shfl_xor_sync(0xffffffffu, hi, o));
+    }
+    const float scale = hi > lo ? (float)PF_NB / (hi - lo) : 0.0f;
+    auto bucket = [&](float v) {
+        if (!(v < INFINITY) || !(v == v)) return PF_NB - 1;
+        const int b = (int)((v - lo) * scale);
+        return b < 0 ? 0 : (b >= PF_NB ? PF_NB - 1 : b);
+    };
+    for (int j = threadIdx.x; j < k; j += blockDim.x) atomicAdd(&cnt[bucket(key(j))], 1u);
+    __syncthreads();
+    // exclusive scan: four buckets a thread, then the warps' and the block's sums
+    unsigned int c4[4], s = 0;
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+        c4[u] = cnt[4 * threadIdx.x + u];
+        s += c4[u];
+    }
+    unsigned int inc = s;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+        const unsigned int t = __shfl_up_sync(0xffffffffu, inc, o);
+        if (lane >= o) inc += t;
+    }
+    __shared__ unsigned int wsum[32];
+    if (lane == 31) wsum[warp] = inc;
+    __syncthreads();
+    if (warp == 0) {
+        unsigned int w = wsum[lane], wi = w;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+            const unsigned int t = __shfl_up_sync(0xffffffffu, wi, o);
+            if (lane >= o) wi += t;
+        }
+        wsum[lane] = wi - w;  // exclusive
+    }
+    __syncthreads();
+    unsigned int run = wsum[warp] + inc - s;
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+        cnt[4 * threadIdx.x + u] = run;
+        run += c4[u];
+    }
+    __syncthreads();
+    for (int j = threadIdx.x; j < k; j += blockDim.x) perm[atomicAdd(&cnt[bucket(key(j))], 1u)] = j;
+}
+
+// The sorted operand rows (F bf16 each), records (||c_F||^2, h') and each
+// 32-position chunk's smallest ||c_F||^2 (positions past k: +inf).  One warp
+// per chunk.
+__global__ void pf_gather_kernel(const uint16_t *__restrict__ cs0, const float4 *__restrict__ cinfo0, int k, int kp,
+                                 int F, const int32_t *__restrict__ perm, uint16_t *__restrict__ cs,
+                                 float4 *__restrict__ cinfo, float *__restrict__ cmin) {
+    const int lane = threadIdx.x & 31;
+    const int64_t w0 = (blockIdx.x * (int64_t)blockDim.x + threadIdx.x) >> 5;
+    const int64_t nw = ((int64_t)gridDim.x * blockDim.x) >> 5;
+    const float *cf0 = reinterpret_cast<const float *>(cinfo0);
+    float *cf = reinterpret_cast<float *>(cinfo);
+    for (int64_t w = w0; w < kp / 32; w += nw) {
+        const int pos = (int)(32 * w) + lane;
+        const int j = pos < k ? perm[pos] : -1;
+        const float cn = j >= 0 ? cf0[4 * (j >> 1) + (j & 1)] : INFINITY;
+        const float h = j >= 0 ? cf0[4 * (j >> 1) + 2 + (j & 1)] : 0.0f;
+        cf[4 * (pos >> 1) + (pos & 1)] = cn;
+        cf[4 * (pos >> 1) + 2 + (pos & 1)] = h;
+        float m = cn;
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) m = fminf(m, __shfl_xor_sync(0xffffffffu, m, o));
+        if (lane == 0) cmin[w] = m;
+        // rows of F bf16 (F % 4 == 0): lanes over 8-byte words
+        for (int r = 0; r < 32; ++r) {
+            const int jr = __shfl_sync(0xffffffffu, j, r);
+            if (jr < 0) break;  // warp-uniform: positions past k are last
+            const uint2 *src = reinterpret_cast<const uint2 *>(cs0 + (int64_t)jr * F);
+            uint2 *dst = reinterpret_cast<uint2 *>(cs + ((int64_t)32 * w + r) * F);
+            for (int q = lane; q < F / 4; q += 32) dst[q] = src[q];
         }
     }
 }
@@ -1827,28 +2077,31 @@ int device_sms() {
 
 template <int MODE, bool SEG, bool PK>
 int launch_tc_kind(const void *xs, int64_t n, int dp, int d, const void *cs, int k, const TcParams &p0,
-                   cudaStream_t st);
+                   cudaStream_t st, int dpb);
 
 // packed: xs is the 1-bit codes [n][ceil(d/32)] or the LVQ4 nibble words
 // [n][ceil(d/8)] (MODE_RBQ1 / MODE_LVQ4)
+// (dpb: the centroid operand's row stride when it differs from dp)
 template <int MODE>
 int launch_tc(const void *xs, int64_t n, int dp, int d, const void *cs, int k, const TcParams &p0,
-              cudaStream_t st, bool packed = false) {
+              cudaStream_t st, bool packed = false, int dpb = -1) {
+    if (dpb < 0) dpb = dp;
     if constexpr (MODE == MODE_RBQ1 || MODE == MODE_LVQ4) {
         if (packed) {
-            if (p0.seg_group) return launch_tc_kind<MODE, true, true>(xs, n, dp, d, cs, k, p0, st);
-            return launch_tc_kind<MODE, false, true>(xs, n, dp, d, cs, k, p0, st);
+            if (p0.seg_group) return launch_tc_kind<MODE, true, true>(xs, n, dp, d, cs, k, p0, st, dpb);
+            return launch_tc_kind<MODE, false, true>(xs, n, dp, d, cs, k, p0, st, dpb);
         }
     }
-    if (p0.seg_group) return launch_tc_kind<MODE, true, false>(xs, n, dp, d, cs, k, p0, st);
-    return launch_tc_kind<MODE, false, false>(xs, n, dp, d, cs, k, p0, st);
+    if constexpr (MODE != MODE_PFRONT)
+        if (p0.seg_group) return launch_tc_kind<MODE, true, false>(xs, n, dp, d, cs, k, p0, st, dpb);
+    return launch_tc_kind<MODE, false, false>(xs, n, dp, d, cs, k, p0, st, dpb);
 }
 
 // One persistent CTA per SM (at most one point tile per CTA when there are
 // fewer tiles than SMs).
 template <int MODE, bool SEG, bool PK>
 int launch_tc_kind(const void *xs, int64_t n, int dp, int d, const void *cs, int k, const TcParams &p0,
-                   cudaStream_t st) {
+                   cudaStream_t st, int dpb) {
     constexpr int NH = TC_NH[MODE];
     constexpr int NS = TC_NS[MODE];
     constexpr size_t SMEM = tc_smem_bytes<MODE, NH, NS>();
@@ -1858,7 +2111,7 @@ int launch_tc_kind(const void *xs, int64_t n, int dp, int d, const void *cs, int
     // the dynamic shared memory attribute, set once per device
     constexpr int MAXDEV = 64;
     static std::mutex mu;
-    static bool attr_set[5][2][2][MAXDEV] = {};
+    static bool attr_set[6][2][2][MAXDEV] = {};
     int dev = 0;
     SKM_CUDA_TRY(cudaGetDevice(&dev));
     {
@@ -1880,7 +2133,7 @@ int launch_tc_kind(const void *xs, int64_t n, int dp, int d, const void *cs, int
     } else {
         SKM_TRY(make_map(&ma, xs, parts * n, d, dp, BM, eb));
     }
-    SKM_TRY(make_map(&mb, cs, (int64_t)parts * k, d, dp, BN, eb));
+    SKM_TRY(make_map(&mb, cs, (int64_t)parts * k, d, dpb, BN, eb));
     TcParams p = p0;
     p.n = n;
     p.nrt = cdiv(n, BM);
@@ -2098,6 +2351,92 @@ void tc_plan(int repr, int64_t n, int d, int k, const void *x, const void *scree
     }
 }
 
+bool tc_pfront_ok(int repr, int d, const void *x) {
+    return repr == SKM_REPR_BF16 && d >= 2 * PF_DIMS && d <= 1024 && d % 8 == 0 && ((uintptr_t)x & 15) == 0;
+}
+
+void tc_plan_pfront(int64_t n, int d, int k, Carver &cv, TcAssignBufs &b) {
+    (void)d;
+    const size_t kp = (size_t)cdiv(k, BN) * BN;
+    b.cs = cv.take<uint16_t>((size_t)k * PF_DIMS);  // sorted by ||c_F||^2
+    b.cinfo = cv.take<float4>(kp / 2);
+    b.cinfoz = cv.take<float2>(kp / 2);
+    b.pf_cs0 = cv.take<uint16_t>((size_t)k * PF_DIMS);  // centroid order
+    b.pf_cinfo0 = cv.take<float4>(kp / 2);
+    b.pf_perm = cv.take<int32_t>(kp);
+    b.pf_cmin = cv.take<float>(kp / 32);
+    b.pf_thr = cv.take<float2>(n);
+    b.pf_cand = cv.take<uint16_t>((size_t)n * PF_CAP);
+    b.pf_cnt = cv.take<int32_t>(n);
+    b.resc_rows = cv.take<int32_t>(n);
+    b.fall_rows = cv.take<int32_t>(n);
+}
+
+// Exact dimension pruning with a tensor-core front (Section 3.1
+// "SuperKMeans": a GEMM over the front dimensions, then pruning on the
+// survivors).  The pruned distance of the method is the fp32 sum of 32-
+// dimension block partials, in order, of (x_i - c_i)^2; a centroid may be
+// dropped once a lower bound of it exceeds the row's seed distance (the
+// distance to its previous centroid), which every argmin and tie is below.
+//   1. centroids: bf16 operand and bound records over the first PF_DIMS
+//      dimensions (the screen's interval terms, with prefix norms);
+//   2. rows: the seed distance and the threshold on s~ over the front
+//      (k_prune.cu);
+//   3. tcgen05 over the front: survivors listed per row; a row whose one
+//      survivor is its seed is decided;
+//   4. CUDA cores: the listed rows' survivors evaluated block by block, and
+//      rows whose lists overflowed pruned over all k.
+// The result is the same as the CUDA-core pruning kernels' bit for bit.
+int tc_assign_pfront(const skm_data *x, const float *C, int k, const int32_t *prev, int32_t *assign, float *dist,
+                     TcAssignBufs &b, unsigned long long *ctr, cudaStream_t st) {
+    const int64_t n = x->n;
+    const int d = x->d;
+    constexpr int F = PF_DIMS;
+    const int kp = (int)(cdiv(k, BN) * BN);
+    SKM_CUDA_TRY(cudaMemsetAsync(b.counters, 0, sizeof(int32_t) * 8, st));
+    const float eps_acc = (float)(((F / BK) * (BK / 16) + 4) * 0x1p-18);
+    const float eps_s = 0x1p-21f;
+    // bf16 points are their own operand: no residual term (counters[7] = 0.0f)
+    cprep_f32_kernel<<<grid_warps(kp), 256, 0, st>>>(C, k, kp, d, F, F, eps_acc, eps_s,
+                                                     reinterpret_cast<const float *>(b.counters + 7),
+                                                     (__nv_bfloat16 *)b.pf_cs0, b.pf_cinfo0, b.cinfoz,
+                                                     reinterpret_cast<unsigned int *>(b.counters + 4), nullptr,
+                                                     nullptr, nullptr, n, nullptr);
+    SKM_CUDA_TRY(launched());
+    // columns sorted by ||c_F||^2 (a chunk's columns then share a tight bound)
+    pf_sort_kernel<<<1, 1024, 0, st>>>(b.pf_cinfo0, k, b.pf_perm);
+    SKM_CUDA_TRY(launched());
+    pf_gather_kernel<<<std::max(1, std::min(kp / 32 / 8, 152 * 8)), 256, 0, st>>>(b.pf_cs0, b.pf_cinfo0, k, kp, F,
+                                                                                  b.pf_perm, b.cs, b.cinfo,
+                                                                                  b.pf_cmin);
+    SKM_CUDA_TRY(launched());
+    const uint16_t *X = static_cast<const uint16_t *>(x->x);
+    SKM_CUDA_TRY(launch_prune_front_prep(X, n, d, F, C, k, prev, reinterpret_cast<const float *>(b.counters + 4),
+                                         b.pf_thr, ctr, st));
+    TcParams p{};
+    p.cinfo = b.cinfo;
+    p.counters = b.counters;
+    p.assign = assign;
+    p.dist = dist;
+    p.resc_rows = b.resc_rows;
+    p.fall_rows = b.fall_rows;
+    p.pf_thr = b.pf_thr;
+    p.pf_cand = b.pf_cand;
+    p.pf_cnt = b.pf_cnt;
+    p.pf_prev = prev;
+    p.pf_ctr = ctr;
+    p.pf_perm = b.pf_perm;
+    p.pf_cmin = b.pf_cmin;
+    SKM_TRY(launch_tc<MODE_PFRONT>(X, n, d, F, b.cs, k, p, st, false, F));
+    constexpr int nsub = TC_NH[MODE_PFRONT] / TC_NS[MODE_PFRONT];
+    SKM_CUDA_TRY(launch_prune_finish(X, d, C, b.pf_thr, b.pf_cand, b.pf_cnt, PF_CAP, nsub, b.pf_perm, b.resc_rows,
+                                     ctr + 4, assign, dist, ctr, st));
+    SKM_CUDA_TRY(launch_prune_rows_cta(X, d, C, k, prev, b.pf_thr, b.fall_rows, ctr + 5, assign, dist, ctr + 6, st));
+    add_stats_kernel<<<1, 1, 0, st>>>(b.counters, b.stats);
+    SKM_CUDA_TRY(launched());
+    return SKM_OK;
+}
+
 int tc_init_stats(TcAssignBufs &b, cudaStream_t st) {
     SKM_CUDA_TRY(cudaMemsetAsync(b.stats, 0, sizeof(int64_t) * 4, st));
     return SKM_OK;
@@ -2139,7 +2478,7 @@ int tc_assign_float(const skm_data *x, const float *C, int k, int32_t *assign, f
     SKM_CUDA_TRY(cudaMemsetAsync(b.counters, 0, sizeof(int32_t) * 8, st));
     // SKM_FLAG_WARM (not in segmented calls): bounds carried between calls
     const bool warm = !seg && (x->flags & SKM_FLAG_WARM) && b.warm_hdr;
-    cprep_f32_kernel<<<grid_warps(kp), 256, 0, st>>>(C, k, kp, d, dp, eps_acc, eps_s, v.rho_max,
+    cprep_f32_kernel<<<grid_warps(kp), 256, 0, st>>>(C, k, kp, d, dp, d, eps_acc, eps_s, v.rho_max,
                                                      (__nv_bfloat16 *)b.cs, b.cinfo, b.cinfoz,
                                                      reinterpret_cast<unsigned int *>(b.counters + 4),
                                                      warm ? b.warm_cprev : nullptr, b.warm_shift, b.warm_hdr, n,

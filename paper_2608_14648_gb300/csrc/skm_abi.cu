@@ -125,8 +125,25 @@ static bool use_prune(const skm_data *x) {
                                           x->repr == SKM_REPR_SQ8 || x->repr == SKM_REPR_RBQ1);
 }
 
+// Pruning counters, the first buffer of every assignment workspace: [0] pairs
+// alive after the first block (or after the tensor-core front), [1]
+// complete, [2] blocks evaluated after the first (the front's finish: every
+// block it evaluated), [3] front dimensions (0: CUDA cores only), [4] rows the
+// front listed for the CUDA-core finish, [5] rows pruned over all k after a
+// list overflow, [6..8] that pruning's own [0..2], [9] k.
+constexpr int PRUNE_CTRS = 10;
+
+static void prune_stats_from(const unsigned long long (&h)[PRUNE_CTRS], skm_stats *out) {
+    out->prune_first_block = (int64_t)h[0];
+    out->prune_complete = (int64_t)(h[1] + h[7]);
+    out->prune_blocks = (int64_t)(h[2] + h[8] + h[5] * h[9]);
+    out->prune_front_dims = (int64_t)h[3];
+    out->prune_rows_finished = (int64_t)h[4];
+    out->prune_rows_full = (int64_t)h[5];
+}
+
 struct AssignBufs {
-    unsigned long long *prune = nullptr;    // [0] pairs alive after block 1, [1] complete, [2] later blocks
+    unsigned long long *prune = nullptr;    // PRUNE_CTRS counters
     int32_t *nx = nullptr, *nc = nullptr;  // SQ8 with d > 1024 (__dp4a path)
     uint4 *planes = nullptr;                // RBQ1 with d > 1024 (AND + popcount path)
     Rbq1CInfo *info = nullptr;
@@ -139,13 +156,15 @@ struct AssignBufs {
 static void plan_assign(const skm_data *x, int k, Carver &cv, AssignBufs &b) {
     const int64_t n = x->n;
     const int d = x->d;
-    b.prune = cv.take<unsigned long long>(3);
+    b.prune = cv.take<unsigned long long>(PRUNE_CTRS);
     if (use_prune(x)) {
         if (x->repr == SKM_REPR_RBQ1) {
             b.planes = cv.take<uint4>((size_t)k * words_of(d));
             b.seginfo = cv.take<Rbq1SegInfo>(k);
         }
         tc_plan(-1, n, d, k, x->x, x->screen, false, cv, b.tc);  // statistics only
+        // bf16 points: the tensor-core front, taken when a seed assignment is given
+        if (tc_pfront_ok(x->repr, d, x->x)) tc_plan_pfront(n, d, k, cv, b.tc);
         return;
     }
     switch (x->repr) {
@@ -270,6 +289,8 @@ static int do_assign(const skm_data *x, const void *C, int k, const int32_t *pre
                                                 b.prune, st));
             return SKM_OK;
         }
+        if (prev && b.tc.pf_thr && tc_pfront_ok(x->repr, d, x->x) && ((uintptr_t)C & 15) == 0)
+            return tc_assign_pfront(x, static_cast<const float *>(C), k, prev, assign, dist, b.tc, b.prune, st);
         if (x->repr == SKM_REPR_SQ8)
             SKM_CUDA_TRY(launch_prune_assign_sq8(static_cast<const uint8_t *>(x->x), n, d, static_cast<const uint8_t *>(C),
                                                  k, prev, assign, dist, b.prune, st));
@@ -755,7 +776,7 @@ int skm_assign(const skm_data *x, const void *C, int k, const int32_t *prev_assi
     plan_assign(x, k, cv, b);
     SKM_TRY(need_ws(cv, ws_bytes, ws));
     if (use_prune(x))
-        SKM_CUDA_TRY(cudaMemsetAsync(b.prune, 0, 3 * sizeof(unsigned long long), S(stream)));
+        SKM_CUDA_TRY(cudaMemsetAsync(b.prune, 0, PRUNE_CTRS * sizeof(unsigned long long), S(stream)));
     return do_assign(x, C, k, prev_assign, assign, dist, b, S(stream));
 }
 
@@ -763,15 +784,13 @@ int skm_assign_prune_stats(const void *ws, size_t ws_bytes, skm_stats *out, void
     if (!ws || !out) return set_error(SKM_ERR_INVALID_ARG, "ws and out are required");
     // the counters are the first buffer of every assignment workspace
     Carver cv(const_cast<void *>(ws), ws_bytes);
-    const unsigned long long *cnt = cv.take<unsigned long long>(3);
+    const unsigned long long *cnt = cv.take<unsigned long long>(PRUNE_CTRS);
     if (!cv.fits()) return set_error(SKM_ERR_INVALID_ARG, "ws_bytes is smaller than the counters");
-    unsigned long long h[3];
+    unsigned long long h[PRUNE_CTRS];
     SKM_CUDA_TRY(cudaMemcpyAsync(h, cnt, sizeof(h), cudaMemcpyDeviceToHost, S(stream)));
     SKM_CUDA_TRY(cudaStreamSynchronize(S(stream)));
     memset(out, 0, sizeof(*out));
-    out->prune_first_block = (int64_t)h[0];
-    out->prune_complete = (int64_t)h[1];
-    out->prune_blocks = (int64_t)h[2];
+    prune_stats_from(h, out);
     return SKM_OK;
 }
 
@@ -1142,7 +1161,7 @@ int skm_fit(const skm_fit_config *cfg, const skm_data *x, const void *C_init,
     // the iterations' screens start from the bounds the previous one left
     if (x->repr == SKM_REPR_F32 || x->repr == SKM_REPR_BF16) xd.flags |= SKM_FLAG_WARM;
     SKM_TRY(tc_init_stats(b.a.tc, st));
-    SKM_CUDA_TRY(cudaMemsetAsync(b.a.prune, 0, 3 * sizeof(unsigned long long), st));
+    SKM_CUDA_TRY(cudaMemsetAsync(b.a.prune, 0, PRUNE_CTRS * sizeof(unsigned long long), st));
     int e = 0;
     if (x->repr == SKM_REPR_RBQ1) {
         SKM_CUDA_TRY(launch_rbq1_exponent(x->F, n, b.maxbits, b.e_dev, st));
@@ -1225,11 +1244,9 @@ int skm_fit(const skm_fit_config *cfg, const skm_data *x, const void *C_init,
     int32_t uflag = 0;
     SKM_CUDA_TRY(cudaMemcpy(&uflag, b.u.flag, sizeof(uflag), cudaMemcpyDeviceToHost));
     if (uflag) return set_error(SKM_ERR_TIMEOUT, "an update pipeline wait exceeded its limit");
-    unsigned long long pr[3] = {0, 0, 0};
+    unsigned long long pr[PRUNE_CTRS] = {};
     SKM_CUDA_TRY(cudaMemcpy(pr, b.a.prune, sizeof(pr), cudaMemcpyDeviceToHost));
-    local.prune_first_block = (int64_t)pr[0];
-    local.prune_complete = (int64_t)pr[1];
-    local.prune_blocks = (int64_t)pr[2];
+    prune_stats_from(pr, &local);
     if (stats_host) {
         int64_t *per_iter = stats_host->empty_per_iter;
         local.empty_per_iter = per_iter;

@@ -40,6 +40,17 @@ struct TcAssignBufs {
     int32_t *resc_rows = nullptr;
     int32_t *fall_rows = nullptr;
     unsigned long long *fall_keys = nullptr;  // F32/BF16: per fallback row, (dist bits, index)
+    // BF16 with SKM_FLAG_PRUNE (tensor-core front): per row (threshold, seed
+    // distance), survivor lists, per listed row the sub-lists' counts
+    float2 *pf_thr = nullptr;
+    uint16_t *pf_cand = nullptr;
+    int32_t *pf_cnt = nullptr;
+    // ... and the centroid operand / records in centroid order (the sorted
+    // copies are cs / cinfo), the sort's permutation and chunk minima
+    uint16_t *pf_cs0 = nullptr;
+    float4 *pf_cinfo0 = nullptr;
+    int32_t *pf_perm = nullptr;
+    float *pf_cmin = nullptr;
 };
 
 // Segmented assignment: rows sorted by group, row r only takes centroids
@@ -61,6 +72,16 @@ bool tc_reads_packed(int repr, int d, const void *x);
 void tc_plan(int repr, int64_t n, int d, int k, const void *x, const void *screen, bool warm, Carver &cv,
              TcAssignBufs &b);
 int tc_init_stats(TcAssignBufs &b, cudaStream_t st);
+// Exact dimension pruning of bf16 points with the first dimensions on tensor
+// cores (used when a seed assignment is given): whether these points can take
+// it, its workspace, and the call.  ctr: the pruning counters ([0] pairs alive
+// after the front, [1] complete, [2] 32-dimension blocks evaluated on CUDA
+// cores, [3] front dimensions, [4] rows finished on CUDA cores, [5] rows
+// pruned over all k, [6..8] the latter's own counters, [9] k).
+bool tc_pfront_ok(int repr, int d, const void *x);
+void tc_plan_pfront(int64_t n, int d, int k, Carver &cv, TcAssignBufs &b);
+int tc_assign_pfront(const skm_data *x, const float *C, int k, const int32_t *prev, int32_t *assign, float *dist,
+                     TcAssignBufs &b, unsigned long long *ctr, cudaStream_t st);
 int tc_assign_float(const skm_data *x, const float *C, int k, int32_t *assign, float *dist,
                     TcAssignBufs &b, cudaStream_t st, const TcSeg *seg = nullptr);
 // nx_plain / nc_plain: buffers for the __dp4a path (d > TC_SQ8_MAX_D), filled here.

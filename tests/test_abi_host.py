@@ -301,3 +301,23 @@ def test_lvq4_packed_reading_needs_no_screen_workspace(skm):
         copied = L.skm_workspace_size(0, ctypes.byref(data(d, 0x1004, n)), 1000)
         assert packed < n * d // 4 and copied >= n * d
     assert L.skm_workspace_size(0, ctypes.byref(data(1000, 0x1000, n)), 1000) >= n * 1000  # 125 words
+
+
+def test_prune_front_workspace_holds_survivor_lists(skm):
+    """bf16 points with SKM_FLAG_PRUNE, 256 <= d <= 1024, d % 8 == 0 and a
+    16-byte aligned base can take the tensor-core front: the workspace then
+    holds the per-row survivor lists (64 int32) and thresholds; other
+    shapes prune on CUDA cores only and need no per-row buffers."""
+    L = skm.lib()
+
+    def data(d, ptr, n):
+        x = skm.Data(skm.REPR_BF16, d, n, ptr, None, None, None, None, 0, 0)
+        x.flags = skm.FLAG_PRUNE
+        return x
+
+    n, k = 100_000, 1000
+    for d in (256, 512, 1024):
+        ws = L.skm_workspace_size(0, ctypes.byref(data(d, 0x1000, n)), k)
+        assert ws >= n * (64 + 5) * 4
+    for d, ptr in ((128, 0x1000), (1032, 0x1000), (260, 0x1000), (256, 0x1008)):
+        assert L.skm_workspace_size(0, ctypes.byref(data(d, ptr, n)), k) < n * 4

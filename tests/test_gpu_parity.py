@@ -545,6 +545,17 @@ def test_prune_assign_vs_oracle_and_seed_independent(skm, repr_name, n, d, k):
     assert torch.equal(d1, d0) and torch.equal(d2, d0)
     nb = (d + 31) // 32
     for st in (st1, st2):
+        if st["prune_front_dims"]:
+            # bf16 with a seed: the tensor-core front screened 128 dimensions
+            # of every pair; every row keeps at least its seed; complete pairs
+            # evaluated all nb blocks on CUDA cores
+            assert repr_name == "bf16" and d >= 256 and st["prune_front_dims"] == 128
+            assert n <= st["prune_first_block"] <= n * k
+            assert 0 <= st["prune_complete"] <= st["prune_first_block"]
+            assert st["prune_rows_finished"] + st["prune_rows_full"] <= n
+            assert st["prune_complete"] * nb <= st["prune_blocks"]
+            assert st["prune_blocks"] <= (st["prune_first_block"] + st["prune_rows_full"] * k) * nb
+            continue
         # every pair evaluates its first block; a pair alive after block b
         # evaluates block b + 1; complete pairs evaluated all nb blocks
         assert 0 < st["prune_complete"] <= st["prune_first_block"] <= n * k
@@ -554,6 +565,55 @@ def test_prune_assign_vs_oracle_and_seed_independent(skm, repr_name, n, d, k):
     # and the tensor-core screen reaches the same assignment
     a3, _ = skm.skm_assign(pts, Cd)
     assert (a3 == a0).float().mean().item() >= AGREE
+
+
+@pytest.mark.parametrize("n,d,k", [(3000, 256, 1000), (1000, 512, 300), (700, 1024, 257), (5000, 256, 13),
+                                   (130, 256, 600)])
+def test_prune_front_tensor_cores_bitexact(skm, n, d, k):
+    """bf16 points with a seed assignment: the first 128 dimensions of every
+    pair screened on tensor cores, survivors finished on CUDA cores (Section
+    3.1 "SuperKMeans", a GEMM over the front dimensions, then pruning).  The
+    result equals the CUDA-core pruning's (seed 0, no front) bit for bit,
+    assignments and distances, with good seeds (most rows decided by the
+    front), in place (seed array = output), and with random seeds (lists
+    overflow to the full pruning); and it matches the oracle."""
+    X = _points(n, d, seed=n + d + k)
+    Xd = X.to(DEV).to(torch.bfloat16).view(torch.int16)
+    xb = Xd.cpu().numpy().view(np.uint16)
+    g = torch.Generator().manual_seed(k)
+    # fp32 centroids off the bf16 grid (the bound's residual terms matter)
+    C = torch.from_numpy(oracle.bf16_to_f32(xb[synth.forgy_indices(n, k, seed=5).numpy()]).copy())
+    C = (C + 0.01 * C.std() * torch.randn(C.shape, generator=g)).contiguous()
+    Cd = C.to(DEV)
+    pp = skm.Points(skm.REPR_BF16, Xd, d, flags=skm.FLAG_PRUNE)
+    a0, d0 = skm.skm_assign(pp, Cd)  # no seed: CUDA cores only
+    a_or, best, second = oracle.assign_bf16(xb, C.numpy())
+    _check_f32(a0.cpu().numpy(), d0.cpu().numpy(), best, second, a_or, f"prune n={n} d={d} k={k}")
+    seed_good, _ = skm.skm_assign(skm.Points(skm.REPR_BF16, Xd, d).with_screen(), Cd)
+    ws = skm.workspace(skm.OP_ASSIGN, pp, k)
+    a1, d1 = skm.skm_assign(pp, Cd, prev_assign=seed_good, ws=ws)
+    st = skm.skm_assign_prune_stats(ws)
+    assert torch.equal(a1, a0) and torch.equal(d1, d0)
+    assert st["prune_front_dims"] == 128
+    assert n <= st["prune_first_block"] <= n * k
+    assert st["prune_rows_finished"] + st["prune_rows_full"] <= n
+    inplace = seed_good.clone()
+    dd = torch.empty(n, device=DEV, dtype=torch.float32)
+    skm.skm_assign(pp, Cd, prev_assign=inplace, ws=ws, out=inplace, dist_out=dd)
+    assert torch.equal(inplace, a0) and torch.equal(dd, d0)
+    seed_bad = torch.randint(0, k, (n,), generator=g, dtype=torch.int32).to(DEV)
+    a2, d2 = skm.skm_assign(pp, Cd, prev_assign=seed_bad, ws=ws)
+    st2 = skm.skm_assign_prune_stats(ws)
+    assert torch.equal(a2, a0) and torch.equal(d2, d0)
+    assert st2["prune_first_block"] >= st["prune_first_block"]
+    if k >= 300:
+        assert st2["prune_rows_full"] > 0  # random seeds keep more than a list holds (128)
+    # without distances, and seeds outside [0, k) (centroid 0)
+    seed_out = seed_good.clone()
+    seed_out[::7] = -1
+    seed_out[3::7] = k
+    a3, _ = skm.skm_assign(pp, Cd, prev_assign=seed_out, ws=ws, want_dist=False)
+    assert torch.equal(a3, a0)
 
 
 @pytest.mark.parametrize("repr_name", ["bf16", "f32"])
