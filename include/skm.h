@@ -107,8 +107,15 @@ enum {
      * pairs far from the nearest are not listed as candidates.  The result
      * is the same; only the work changes.  A workspace whose last call had
      * other n, d or k, or did not finish, starts cold.  The caller must not
-     * change the points between such calls.  skm_fit uses it between its
-     * iterations. */
+     * change the points between such calls, and a workspace first used with
+     * this flag must be zero-filled (or come from a call on these points).
+     * skm_fit uses it between its iterations (clearing it first).
+     * BF16 with SKM_FLAG_PRUNE and the tensor-core front (see skm_assign): each
+     * row keeps an upper bound U of its pruned distance to its centroid; the
+     * next call grows it by the centroid's move, U' = (sqrt(U (1 + g)) +
+     * ||c' - c||)^2 (1 + g) with g covering the fp32 rounding, and forms the
+     * front's threshold from U' without reading the points.  Calls that want
+     * distances use the exact seed distances instead. */
     SKM_FLAG_WARM = 4
 };
 

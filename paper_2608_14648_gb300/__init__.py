@@ -181,10 +181,12 @@ def _stream(stream=None):
     return ctypes.c_void_p(s.cuda_stream)
 
 
-def _ws(nbytes, device):
+def _ws(nbytes, device, zero=False):
     nbytes = max(int(nbytes), 256)
-    # 256-byte alignment: the caching allocator returns 512-byte aligned blocks
-    return torch.empty(nbytes, dtype=torch.uint8, device=device)
+    # 256-byte alignment: the caching allocator returns 512-byte aligned blocks;
+    # zero: a workspace that carries state between calls (SKM_FLAG_WARM) starts
+    # with no stamp, whatever the recycled memory held
+    return (torch.zeros if zero else torch.empty)(nbytes, dtype=torch.uint8, device=device)
 
 
 def _dev(t):
@@ -394,8 +396,10 @@ def skm_rbq1_exponent(F, stream=None):
 
 
 def workspace(op, pts: Points, k):
-    """A device workspace tensor sized for op (OP_ASSIGN, OP_UPDATE, OP_FIT)."""
-    return _ws(skm_workspace_size(op, pts, k), pts.device)
+    """A device workspace tensor sized for op (OP_ASSIGN, OP_UPDATE, OP_FIT),
+    zero-filled (a workspace that carries bounds between calls must start
+    without a stamp)."""
+    return _ws(skm_workspace_size(op, pts, k), pts.device, zero=True)
 
 
 def rbq1_points(q, d, e=None):
@@ -595,7 +599,7 @@ class LloydStepHost:
         nbytes = lib().skm_step_host_workspace_size(ctypes.byref(self.cfg), ctypes.byref(self.ref))
         if nbytes == 0:
             raise SkmError(1, lib().skm_last_error().decode())
-        self.ws = _ws(nbytes, self.device)
+        self.ws = _ws(nbytes, self.device, zero=True)
 
     def _exchange(self, partial, counts, user, stream):
         # the hook's work goes on the stream this step was called with (the

@@ -191,9 +191,10 @@ __global__ void __launch_bounds__(PR_WARPS * 32) prune_assign_kernel(
 // CTA keeps the smallest (distance, index) of the warps' results.
 constexpr int PRC_WARPS = 8;
 __global__ void __launch_bounds__(PRC_WARPS * 32) prune_rows_cta_kernel(
-    const uint16_t *__restrict__ X, int d, const float *__restrict__ C, int k, const int32_t *__restrict__ prev,
-    const float2 *__restrict__ thr, const int32_t *__restrict__ rows, const unsigned long long *__restrict__ nrows,
-    int32_t *__restrict__ assign, float *__restrict__ dist, unsigned long long *__restrict__ counters) {
+    const uint16_t *__restrict__ X, int d, const float *__restrict__ C, int k, const int32_t *__restrict__ seeds,
+    const float2 *__restrict__ thr, int2 *__restrict__ wrow, const int32_t *__restrict__ rows,
+    const int32_t *__restrict__ nrows, int32_t *__restrict__ assign, float *__restrict__ dist,
+    unsigned long long *__restrict__ counters) {
     __shared__ float sx[PR_MAX_D];
     __shared__ int qid[PRC_WARPS][2][PR_BATCH];
     __shared__ float qps[PRC_WARPS][2][PR_BATCH];
@@ -208,8 +209,9 @@ __global__ void __launch_bounds__(PRC_WARPS * 32) prune_rows_cta_kernel(
         __syncthreads();  // the previous row's sx and results are read
         for (int i = threadIdx.x; i < d; i += blockDim.x) sx[i] = ldx<uint16_t>(X + row * d + i);
         __syncthreads();
-        int best = prev ? prev[row] : 0;
-        if (best < 0 || best >= k) best = 0;
+        // the seed and its distance, or an upper bound of it (kept bounds): the
+        // seed itself then completes below it, so the result is the same
+        int best = seeds[row];
         float beta = thr[row].y;
         prune_batches(sx, C, d, k, warp * PR_BATCH, PRC_WARPS * PR_BATCH, slack, beta, best, qid[warp], qps[warp],
                       first_alive, complete, later);
@@ -228,6 +230,7 @@ __global__ void __launch_bounds__(PRC_WARPS * 32) prune_rows_cta_kernel(
                 }
             assign[row] = bj;
             if (dist) dist[row] = bp;
+            if (wrow) wrow[row] = make_int2(__float_as_int(bp), bj);
         }
     }
     if (lane == 0 && (first_alive | complete | later)) {
@@ -604,10 +607,20 @@ __device__ __forceinline__ float block_bf16(const uint16_t *xr, const float *cr,
     return part;
 }
 
+//
+// Kept bounds (the state a previous call on these points left, when its stamp
+// matches and no distances are wanted): the row's bound U >= D(x, c) for its
+// centroid c grows by that centroid's move delta = ||c' - c|| (rounded up).
+// With g = (40 + blocks) 2^-23 (twice the rounding of a pruned distance in
+// either direction), the real squared distance is at most U (1 + g), its root
+// grows by at most delta (triangle inequality), and the new pruned distance
+// is at most U' = (sqrt(U (1 + g)) + delta)^2 (1 + g), every step rounded up;
+// the threshold is then formed from U' as above, with the kept prefix norms.
 __global__ void front_prep_kernel(const uint16_t *__restrict__ X, int64_t n, int d, int F, int G,
                                   const float *__restrict__ C, int k, const int32_t *__restrict__ prev,
-                                  const float *__restrict__ hz, float2 *__restrict__ thr,
+                                  const float *__restrict__ hz, PfRows r, int force_cold,
                                   unsigned long long *__restrict__ ctr) {
+    float2 *__restrict__ thr = r.thr;
     const int lane = threadIdx.x & 31;
     const int sub = lane / G, b = lane % G;
     const int rpw = 32 / G;  // rows per warp
@@ -621,6 +634,28 @@ __global__ void front_prep_kernel(const uint16_t *__restrict__ X, int64_t n, int
     const float H = __ldg(hz), Z = __ldg(hz + 1);
     const float slack = prune_slack(d);
     const float K1 = __fmul_ru(slack, 1.0f + 0x1p-16f);
+    if (r.warm_ok && *r.warm_ok && !force_cold) {
+        const float g = (float)(40 + nb) * 0x1p-23f;
+        const int64_t nt = (int64_t)gridDim.x * blockDim.x;
+        for (int64_t row = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; row < n; row += nt) {
+            const int2 w = r.wrow[row];
+            const float U = __int_as_float(w.x);
+            float t = INFINITY, Un = INFINITY;
+            int seed = 0;
+            if (w.y >= 0 && w.y < k && U >= 0.0f && U < INFINITY) {
+                seed = w.y;
+                const float rr = __fadd_ru(__fsqrt_ru(__fmul_ru(U, 1.0f + g)), __ldg(&r.shift[seed].y));
+                Un = __fmul_ru(__fmul_ru(rr, rr), 1.0f + g);
+                const float2 xn = r.xn[row];
+                const float W = __fmaf_ru(2.0f * xn.x, H, Z);
+                t = __fadd_ru(__fadd_ru(__fsub_ru(__fmul_ru(Un, K1), xn.y), W), 0x1p-100f);
+                if (!(t == t) || !(Un < INFINITY)) t = INFINITY;
+            }
+            thr[row] = make_float2(t, Un);
+            r.seed[row] = seed;
+        }
+        return;
+    }
     for (int64_t r0 = warp * rpw; r0 < n; r0 += nw * rpw) {
         const int64_t row = r0 + sub;
         const bool act = row < n;
@@ -644,6 +679,8 @@ __global__ void front_prep_kernel(const uint16_t *__restrict__ X, int64_t n, int
             t = __fadd_ru(t, 0x1p-100f);
             if (!(t == t) || !(beta0 < INFINITY)) t = INFINITY;
             thr[row] = make_float2(t, beta0);
+            r.seed[row] = seed;
+            if (r.xn) r.xn[row] = make_float2(xn_up, xn2_lo);
         }
     }
 }
@@ -659,8 +696,8 @@ __global__ void front_prep_kernel(const uint16_t *__restrict__ X, int64_t n, int
 __global__ void __launch_bounds__(256) prune_finish_kernel(
     const uint16_t *__restrict__ X, int d, int G, const float *__restrict__ C, const float2 *__restrict__ thr,
     const uint16_t *__restrict__ cand, const int32_t *__restrict__ cnt, int cap, int nsub,
-    const int32_t *__restrict__ perm, const int32_t *__restrict__ rows, const unsigned long long *__restrict__ nrows,
-    int32_t *__restrict__ assign, float *__restrict__ dist, unsigned long long *__restrict__ ctr) {
+    const int32_t *__restrict__ perm, const int32_t *__restrict__ rows, const int32_t *__restrict__ nrows,
+    int32_t *__restrict__ assign, float *__restrict__ dist, int2 *__restrict__ wrow, unsigned long long *__restrict__ ctr) {
     const int lane = threadIdx.x & 31;
     const int slot = lane / G, b = lane % G, S = 32 / G;
     const int nb = (d + 31) >> 5;
@@ -725,6 +762,7 @@ __global__ void __launch_bounds__(256) prune_finish_kernel(
         if (lane == 0) {
             assign[row] = bj;
             if (dist) dist[row] = bp;
+            if (wrow) wrow[row] = make_int2(__float_as_int(bp), bj);
         }
     }
 #pragma unroll
@@ -783,18 +821,18 @@ cudaError_t launch_prune_assign(const void *X, int x_is_bf16, int64_t n, int d, 
     return launched();
 }
 
-cudaError_t launch_prune_rows_cta(const uint16_t *X, int d, const float *C, int k, const int32_t *prev,
-                                  const float2 *thr, const int32_t *rows, const unsigned long long *nrows,
-                                  int32_t *assign, float *dist, unsigned long long *counters, cudaStream_t st) {
+cudaError_t launch_prune_rows_cta(const uint16_t *X, int d, const float *C, int k, const PfRows &r,
+                                  const int32_t *rows, const int32_t *nrows, int32_t *assign,
+                                  float *dist, unsigned long long *counters, cudaStream_t st) {
     if (d > PR_MAX_D) return cudaErrorInvalidValue;
-    prune_rows_cta_kernel<<<152 * 4, PRC_WARPS * 32, 0, st>>>(X, d, C, k, prev, thr, rows, nrows, assign, dist,
-                                                              counters);
+    prune_rows_cta_kernel<<<152 * 4, PRC_WARPS * 32, 0, st>>>(X, d, C, k, r.seed, r.thr, r.wrow, rows, nrows, assign,
+                                                              dist, counters);
     return launched();
 }
 
 cudaError_t launch_prune_front_prep(const uint16_t *X, int64_t n, int d, int F, const float *C, int k,
-                                    const int32_t *prev, const float *hz, float2 *thr, unsigned long long *ctr,
-                                    cudaStream_t st) {
+                                    const int32_t *prev, const float *hz, const PfRows &r, int force_cold,
+                                    unsigned long long *ctr, cudaStream_t st) {
     const int nb = (d + 31) >> 5;
     int G = 1;
     while (G < nb) G <<= 1;
@@ -803,13 +841,13 @@ cudaError_t launch_prune_front_prep(const uint16_t *X, int64_t n, int d, int F, 
     int64_t blocks = (n + per_block - 1) / per_block;
     if (blocks > 152 * 16) blocks = 152 * 16;
     if (blocks < 1) blocks = 1;
-    front_prep_kernel<<<(int)blocks, 256, 0, st>>>(X, n, d, F, G, C, k, prev, hz, thr, ctr);
+    front_prep_kernel<<<(int)blocks, 256, 0, st>>>(X, n, d, F, G, C, k, prev, hz, r, force_cold, ctr);
     return launched();
 }
 
 cudaError_t launch_prune_finish(const uint16_t *X, int d, const float *C, const float2 *thr, const uint16_t *cand,
                                 const int32_t *cnt, int cap, int nsub, const int32_t *perm, const int32_t *rows,
-                                const unsigned long long *nrows, int32_t *assign, float *dist,
+                                const int32_t *nrows, int32_t *assign, float *dist, int2 *wrow,
                                 unsigned long long *ctr, cudaStream_t st) {
     const int nb = (d + 31) >> 5;
     int G = 1;
@@ -817,7 +855,7 @@ cudaError_t launch_prune_finish(const uint16_t *X, int d, const float *C, const 
     if (G > 32 || (d % 8) != 0 || nsub < 1 || nsub > 4 || cap % nsub != 0 || cap / nsub > 255)
         return cudaErrorInvalidValue;
     prune_finish_kernel<<<152 * 8, 256, 0, st>>>(X, d, G, C, thr, cand, cnt, cap, nsub, perm, rows, nrows, assign,
-                                                 dist, ctr);
+                                                 dist, wrow, ctr);
     return launched();
 }
 

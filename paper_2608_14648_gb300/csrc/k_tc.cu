@@ -39,6 +39,7 @@
 #include <cuda.h>
 #include <cudaTypedefs.h>
 
+#include <cfloat>
 #include <mutex>
 
 #include "skm_tc.cuh"
@@ -188,8 +189,9 @@ struct TcParams {
     // pruned distance), survivor lists [n][PF_CAP] (sorted positions, one
     // sub-list of PF_CAP / NHG per column slice), per listed row the
     // sub-lists' counts (8 bits each), the seed centroids (NULL: centroid 0)
-    // and the pruning counters ([0] pairs alive after the front, [4] rows
-    // listed for the CUDA-core finish, [5] rows whose lists overflowed)
+    // and the pruning counters ([0] pairs alive after the front); the rows
+    // listed for the CUDA-core finish and the rows whose lists overflowed
+    // go to resc_rows / fall_rows (counts: counters[0] / counters[1], per call)
     const float2 *pf_thr;
     uint16_t *pf_cand;
     // PFRONT: the centroid operand and records are sorted by ||c_F||^2
@@ -198,8 +200,9 @@ struct TcParams {
     const int32_t *pf_perm;
     const float *pf_cmin;
     int32_t *pf_cnt;
-    const int32_t *pf_prev;
+    const int32_t *pf_seed;
     unsigned long long *pf_ctr;
+    int2 *pf_wrow;  // kept bounds: (bound bits, centroid) of decided rows (NULL: none)
     // Fault injection (0 = off): the producer first waits this long on a
     // barrier that nothing arrives on, so the launch gives up before it has
     // loaded anything and reports through the abort flag.
@@ -957,7 +960,8 @@ __global__ void __launch_bounds__(tc_threads<NH, PK>(), 1)
             int pcnt = 0;
             uint16_t *pf_list = nullptr;
             if (MODE == MODE_PFRONT && valid) {
-                pthr = p.pf_thr[row].x;
+                // finite, so that columns past k (s~ = +inf) never survive
+                pthr = fminf(p.pf_thr[row].x, FLT_MAX);
                 pf_list = p.pf_cand + row * PF_CAP + slice * PF_SUB;
             }
             // segmented mode: this row's centroid range (ids clamped into bounds)
@@ -1368,16 +1372,17 @@ __global__ void __launch_bounds__(tc_threads<NH, PK>(), 1)
                     packed |= (uint32_t)min(ch, 255) << (8 * h);
                 }
                 pf_alive += (unsigned long long)tot;
-                int seed = p.pf_prev ? p.pf_prev[row] : 0;
-                seed = (seed < 0 || seed >= p.k) ? 0 : seed;
+                const int seed = p.pf_seed[row];
                 if (!over && tot == 1 && one >= 0 && p.pf_perm[p.pf_cand[row * PF_CAP + one * PF_SUB]] == seed) {
                     p.assign[row] = seed;
-                    if (p.dist) p.dist[row] = p.pf_thr[row].y;
+                    const float u = p.pf_thr[row].y;  // the seed's distance (or, kept bounds, a bound of it)
+                    if (p.dist) p.dist[row] = u;
+                    if (p.pf_wrow) p.pf_wrow[row] = make_int2(__float_as_int(u), seed);
                 } else if (!over && tot >= 2) {
                     p.pf_cnt[row] = (int32_t)packed;
-                    p.resc_rows[atomicAdd(p.pf_ctr + 4, 1ull)] = (int32_t)row;
+                    p.resc_rows[atomicAdd(p.counters, 1)] = (int32_t)row;
                 } else {
-                    p.fall_rows[atomicAdd(p.pf_ctr + 5, 1ull)] = (int32_t)row;
+                    p.fall_rows[atomicAdd(p.counters + 1, 1)] = (int32_t)row;
                 }
             }
             if (MODE != MODE_PFRONT && slice == 0 && valid && !dead) {
@@ -1697,7 +1702,7 @@ __global__ void cprep_f32_kernel(const float *__restrict__ C, int k, int kp, int
 // order within a bucket is whatever the atomics give: the survivors' lists
 // then differ in order only, which the argmin does not see).
 constexpr int PF_NB = 4096;
-__global__ void __launch_bounds__(1024) pf_sort_kernel(const float4 *__restrict__ cinfo, int k,
+__global__ void __launch_bounds__(1024) pf_sort_kernel(const float4 *__restrict__ cinfo, int k, int kp,
                                                        int32_t *__restrict__ perm) {
     __shared__ unsigned int cnt[PF_NB];
     __shared__ float red[2][32];
@@ -1772,6 +1777,7 @@ __global__ void __launch_bounds__(1024) pf_sort_kernel(const float4 *__restrict_
     }
     __syncthreads();
     for (int j = threadIdx.x; j < k; j += blockDim.x) perm[atomicAdd(&cnt[bucket(key(j))], 1u)] = j;
+    for (int pos = k + threadIdx.x; pos < kp; pos += blockDim.x) perm[pos] = 0;  // padding: a valid index
 }
 
 // The sorted operand rows (F bf16 each), records (||c_F||^2, h') and each
@@ -2355,9 +2361,16 @@ bool tc_pfront_ok(int repr, int d, const void *x) {
     return repr == SKM_REPR_BF16 && d >= 2 * PF_DIMS && d <= 1024 && d % 8 == 0 && ((uintptr_t)x & 15) == 0;
 }
 
-void tc_plan_pfront(int64_t n, int d, int k, Carver &cv, TcAssignBufs &b) {
-    (void)d;
+void tc_plan_pfront(int64_t n, int d, int k, bool warm, Carver &cv, TcAssignBufs &b) {
     const size_t kp = (size_t)cdiv(k, BN) * BN;
+    b.pf_seed = cv.take<int32_t>(n);
+    if (warm) {  // bounds kept across calls
+        b.pf_whdr = cv.take<int64_t>(4);
+        b.pf_wrow = cv.take<int2>(n);
+        b.pf_xn = cv.take<float2>(n);
+        b.pf_cprev = cv.take<float>((size_t)k * d);
+        b.pf_shift = cv.take<float2>(k);
+    }
     b.cs = cv.take<uint16_t>((size_t)k * PF_DIMS);  // sorted by ||c_F||^2
     b.cinfo = cv.take<float4>(kp / 2);
     b.cinfoz = cv.take<float2>(kp / 2);
@@ -2387,8 +2400,28 @@ void tc_plan_pfront(int64_t n, int d, int k, Carver &cv, TcAssignBufs &b) {
 //   4. CUDA cores: the listed rows' survivors evaluated block by block, and
 //      rows whose lists overflowed pruned over all k.
 // The result is the same as the CUDA-core pruning kernels' bit for bit.
+// End of a front call: the call's list counts into the pruning statistics
+// ([4] finished rows, [5] rows pruned over all k; cumulative in skm_fit) and,
+// with kept bounds (hdr), the stamp when no wait gave up (every row's bound
+// was then written).
+__global__ void pf_done_kernel(int64_t *__restrict__ hdr, const int32_t *__restrict__ counters,
+                               unsigned long long *__restrict__ ctr, int64_t n, int d, int k) {
+    ctr[4] += (unsigned long long)counters[0];
+    ctr[5] += (unsigned long long)counters[1];
+    if (hdr && counters[2] == 0) {
+        hdr[1] = n;
+        hdr[2] = d;
+        hdr[3] = k;
+        __threadfence();
+        hdr[0] = WARM_MAGIC;
+    }
+}
+
 int tc_assign_pfront(const skm_data *x, const float *C, int k, const int32_t *prev, int32_t *assign, float *dist,
                      TcAssignBufs &b, unsigned long long *ctr, cudaStream_t st) {
+    // SKM_FLAG_WARM: bounds kept across calls (the previous call's state applies
+    // when its stamp matches; distances wanted: exact seed distances this call)
+    const bool warm = (x->flags & SKM_FLAG_WARM) && b.pf_whdr;
     const int64_t n = x->n;
     const int d = x->d;
     constexpr int F = PF_DIMS;
@@ -2400,19 +2433,29 @@ int tc_assign_pfront(const skm_data *x, const float *C, int k, const int32_t *pr
     cprep_f32_kernel<<<grid_warps(kp), 256, 0, st>>>(C, k, kp, d, F, F, eps_acc, eps_s,
                                                      reinterpret_cast<const float *>(b.counters + 7),
                                                      (__nv_bfloat16 *)b.pf_cs0, b.pf_cinfo0, b.cinfoz,
-                                                     reinterpret_cast<unsigned int *>(b.counters + 4), nullptr,
-                                                     nullptr, nullptr, n, nullptr);
+                                                     reinterpret_cast<unsigned int *>(b.counters + 4),
+                                                     warm ? b.pf_cprev : nullptr, b.pf_shift, b.pf_whdr, n,
+                                                     b.counters + 6);
     SKM_CUDA_TRY(launched());
     // columns sorted by ||c_F||^2 (a chunk's columns then share a tight bound)
-    pf_sort_kernel<<<1, 1024, 0, st>>>(b.pf_cinfo0, k, b.pf_perm);
+    pf_sort_kernel<<<1, 1024, 0, st>>>(b.pf_cinfo0, k, kp, b.pf_perm);
     SKM_CUDA_TRY(launched());
     pf_gather_kernel<<<std::max(1, std::min(kp / 32 / 8, 152 * 8)), 256, 0, st>>>(b.pf_cs0, b.pf_cinfo0, k, kp, F,
                                                                                   b.pf_perm, b.cs, b.cinfo,
                                                                                   b.pf_cmin);
     SKM_CUDA_TRY(launched());
     const uint16_t *X = static_cast<const uint16_t *>(x->x);
+    PfRows rows;
+    rows.thr = b.pf_thr;
+    rows.seed = b.pf_seed;
+    if (warm) {
+        rows.xn = b.pf_xn;
+        rows.wrow = b.pf_wrow;
+        rows.shift = b.pf_shift;
+        rows.warm_ok = b.counters + 6;
+    }
     SKM_CUDA_TRY(launch_prune_front_prep(X, n, d, F, C, k, prev, reinterpret_cast<const float *>(b.counters + 4),
-                                         b.pf_thr, ctr, st));
+                                         rows, dist != nullptr, ctr, st));
     TcParams p{};
     p.cinfo = b.cinfo;
     p.counters = b.counters;
@@ -2423,16 +2466,19 @@ int tc_assign_pfront(const skm_data *x, const float *C, int k, const int32_t *pr
     p.pf_thr = b.pf_thr;
     p.pf_cand = b.pf_cand;
     p.pf_cnt = b.pf_cnt;
-    p.pf_prev = prev;
+    p.pf_seed = b.pf_seed;
     p.pf_ctr = ctr;
+    p.pf_wrow = rows.wrow;
     p.pf_perm = b.pf_perm;
     p.pf_cmin = b.pf_cmin;
     SKM_TRY(launch_tc<MODE_PFRONT>(X, n, d, F, b.cs, k, p, st, false, F));
     constexpr int nsub = TC_NH[MODE_PFRONT] / TC_NS[MODE_PFRONT];
     SKM_CUDA_TRY(launch_prune_finish(X, d, C, b.pf_thr, b.pf_cand, b.pf_cnt, PF_CAP, nsub, b.pf_perm, b.resc_rows,
-                                     ctr + 4, assign, dist, ctr, st));
-    SKM_CUDA_TRY(launch_prune_rows_cta(X, d, C, k, prev, b.pf_thr, b.fall_rows, ctr + 5, assign, dist, ctr + 6, st));
+                                     b.counters, assign, dist, rows.wrow, ctr, st));
+    SKM_CUDA_TRY(launch_prune_rows_cta(X, d, C, k, rows, b.fall_rows, b.counters + 1, assign, dist, ctr + 6, st));
     add_stats_kernel<<<1, 1, 0, st>>>(b.counters, b.stats);
+    SKM_CUDA_TRY(launched());
+    pf_done_kernel<<<1, 1, 0, st>>>(warm ? b.pf_whdr : nullptr, b.counters, ctr, n, d, k);
     SKM_CUDA_TRY(launched());
     return SKM_OK;
 }

@@ -164,7 +164,7 @@ static void plan_assign(const skm_data *x, int k, Carver &cv, AssignBufs &b) {
         }
         tc_plan(-1, n, d, k, x->x, x->screen, false, cv, b.tc);  // statistics only
         // bf16 points: the tensor-core front, taken when a seed assignment is given
-        if (tc_pfront_ok(x->repr, d, x->x)) tc_plan_pfront(n, d, k, cv, b.tc);
+        if (tc_pfront_ok(x->repr, d, x->x)) tc_plan_pfront(n, d, k, (x->flags & SKM_FLAG_WARM) != 0, cv, b.tc);
         return;
     }
     switch (x->repr) {
@@ -1158,8 +1158,11 @@ int skm_fit(const skm_fit_config *cfg, const skm_data *x, const void *C_init,
         SKM_TRY(tc_screen_prep(x, b.screen, st));
         xd.screen = b.screen;
     }
-    // the iterations' screens start from the bounds the previous one left
+    // the iterations' screens start from the bounds the previous one left; the
+    // first starts cold whatever state the workspace held (other points)
     if (x->repr == SKM_REPR_F32 || x->repr == SKM_REPR_BF16) xd.flags |= SKM_FLAG_WARM;
+    if (b.a.tc.warm_hdr) SKM_CUDA_TRY(cudaMemsetAsync(b.a.tc.warm_hdr, 0, 4 * sizeof(int64_t), st));
+    if (b.a.tc.pf_whdr) SKM_CUDA_TRY(cudaMemsetAsync(b.a.tc.pf_whdr, 0, 4 * sizeof(int64_t), st));
     SKM_TRY(tc_init_stats(b.a.tc, st));
     SKM_CUDA_TRY(cudaMemsetAsync(b.a.prune, 0, PRUNE_CTRS * sizeof(unsigned long long), st));
     int e = 0;

@@ -214,24 +214,41 @@ cudaError_t launch_prune_assign(const void *X, int x_is_bf16, int64_t n, int d, 
                                 unsigned long long *counters, cudaStream_t st);
 cudaError_t launch_prune_assign_sq8(const uint8_t *X, int64_t n, int d, const uint8_t *C, int k, const int32_t *prev,
                                     int32_t *assign, float *dist, unsigned long long *counters, cudaStream_t st);
+// Per-row state of the tensor-core pruning front (bf16 points): (threshold
+// on s~ over the front, the seed's pruned distance or an upper bound of it),
+// the seed centroid; with bounds kept across calls (all NULL otherwise):
+// (||x_F|| rounded up, ||x_F||^2 rounded down), (bound bits, centroid) for
+// the next call, per centroid (., ||c' - c||) since the bounds were written,
+// and the device flag saying whether the kept bounds apply.
+struct PfRows {
+    float2 *thr = nullptr;
+    int32_t *seed = nullptr;
+    float2 *xn = nullptr;
+    int2 *wrow = nullptr;
+    const float2 *shift = nullptr;
+    const int32_t *warm_ok = nullptr;
+};
 // the same pruning of bf16 points over the rows rows[0 .. *nrows) only
-// (device count), one CTA per row, from the seed distances thr[row].y
-cudaError_t launch_prune_rows_cta(const uint16_t *X, int d, const float *C, int k, const int32_t *prev,
-                                  const float2 *thr, const int32_t *rows, const unsigned long long *nrows,
-                                  int32_t *assign, float *dist, unsigned long long *counters, cudaStream_t st);
-// Tensor-core pruning front (bf16 points, d <= 1024): per row the pruned
-// distance to its seed centroid and the threshold on s~ over the first F
-// dimensions; hz = (max h', max z) of the front's centroid records.
+// (device count), one CTA per row, from the seeds and distances (or bounds)
+// of r; writes r.wrow when kept
+cudaError_t launch_prune_rows_cta(const uint16_t *X, int d, const float *C, int k, const PfRows &r,
+                                  const int32_t *rows, const int32_t *nrows, int32_t *assign,
+                                  float *dist, unsigned long long *counters, cudaStream_t st);
+// Tensor-core pruning front (bf16 points, d <= 1024): per row the seed, the
+// pruned distance to it and the threshold on s~ over the first F dimensions
+// (hz = (max h', max z) of the front's centroid records); with kept bounds
+// that apply and force_cold == 0, the seed and a bound from the kept state
+// instead, without reading the points.
 cudaError_t launch_prune_front_prep(const uint16_t *X, int64_t n, int d, int F, const float *C, int k,
-                                    const int32_t *prev, const float *hz, float2 *thr, unsigned long long *ctr,
-                                    cudaStream_t st);
+                                    const int32_t *prev, const float *hz, const PfRows &r, int force_cold,
+                                    unsigned long long *ctr, cudaStream_t st);
 // Rows rows[0 .. *nrows) with front survivors cand[row][cap] (nsub sub-lists
 // of cap / nsub, 8-bit counts in cnt[row]; entries are positions, perm[pos]
 // the centroid): the pruned distances of the survivors and the smallest
 // (lowest index on ties).
 cudaError_t launch_prune_finish(const uint16_t *X, int d, const float *C, const float2 *thr, const uint16_t *cand,
                                 const int32_t *cnt, int cap, int nsub, const int32_t *perm, const int32_t *rows,
-                                const unsigned long long *nrows, int32_t *assign, float *dist,
+                                const int32_t *nrows, int32_t *assign, float *dist, int2 *wrow,
                                 unsigned long long *ctr, cudaStream_t st);
 cudaError_t launch_assign_sq8_simt(const uint8_t *X, int64_t n, int d, const uint8_t *C, int k,
                                    const int32_t *nx, const int32_t *nc, int32_t *assign,

@@ -51,6 +51,14 @@ struct TcAssignBufs {
     float4 *pf_cinfo0 = nullptr;
     int32_t *pf_perm = nullptr;
     float *pf_cmin = nullptr;
+    int32_t *pf_seed = nullptr;  // per row: the seed centroid
+    // ... with SKM_FLAG_WARM: stamp, per row (bound bits, centroid) and the
+    // prefix norms, the previous centroids and their moves
+    int64_t *pf_whdr = nullptr;
+    int2 *pf_wrow = nullptr;
+    float2 *pf_xn = nullptr;
+    float *pf_cprev = nullptr;
+    float2 *pf_shift = nullptr;
 };
 
 // Segmented assignment: rows sorted by group, row r only takes centroids
@@ -79,7 +87,7 @@ int tc_init_stats(TcAssignBufs &b, cudaStream_t st);
 // cores, [3] front dimensions, [4] rows finished on CUDA cores, [5] rows
 // pruned over all k, [6..8] the latter's own counters, [9] k).
 bool tc_pfront_ok(int repr, int d, const void *x);
-void tc_plan_pfront(int64_t n, int d, int k, Carver &cv, TcAssignBufs &b);
+void tc_plan_pfront(int64_t n, int d, int k, bool warm, Carver &cv, TcAssignBufs &b);
 int tc_assign_pfront(const skm_data *x, const float *C, int k, const int32_t *prev, int32_t *assign, float *dist,
                      TcAssignBufs &b, unsigned long long *ctr, cudaStream_t st);
 int tc_assign_float(const skm_data *x, const float *C, int k, int32_t *assign, float *dist,

@@ -616,6 +616,50 @@ def test_prune_front_tensor_cores_bitexact(skm, n, d, k):
     assert torch.equal(a3, a0)
 
 
+def test_prune_front_kept_bounds_across_lloyd_steps(skm):
+    """SKM_FLAG_WARM with the tensor-core pruning front: after the first call
+    each row's threshold comes from the bound the previous call left, grown
+    by its centroid's move, without reading the points.  Every Lloyd step's
+    assignment equals the CUDA-core pruning's bit for bit; a call that wants
+    distances gets the exact ones and keeps the state usable; a workspace
+    holding another point set's state (same shapes) is cleared by skm_fit."""
+    n, d, k = 4000, 256, 300
+    X = _points(n, d, seed=77)
+    Xd = X.to(DEV).to(torch.bfloat16).view(torch.int16)
+    xb = Xd.cpu().numpy().view(np.uint16)
+    C = torch.from_numpy(oracle.bf16_to_f32(xb[synth.forgy_indices(n, k, seed=9).numpy()]).copy()).to(DEV)
+    pw = skm.Points(skm.REPR_BF16, Xd, d, flags=skm.FLAG_PRUNE | skm.FLAG_WARM)
+    pc = skm.Points(skm.REPR_BF16, Xd, d, flags=skm.FLAG_PRUNE)
+    ws = skm.workspace(skm.OP_ASSIGN, pw, k)
+    a_prev, _ = skm.skm_assign(pc, C)  # no seed: CUDA cores
+    for it in range(6):
+        a_c, d_c = skm.skm_assign(pc, C)
+        if it == 3:  # distances wanted: exact seed distances this call
+            a_w, d_w = skm.skm_assign(pw, C, prev_assign=a_prev, ws=ws)
+            assert torch.equal(d_w, d_c)
+        else:
+            a_w, _ = skm.skm_assign(pw, C, prev_assign=a_prev, ws=ws, want_dist=False)
+        assert torch.equal(a_w, a_c), f"step {it}"
+        st = skm.skm_assign_prune_stats(ws)
+        assert st["prune_front_dims"] == 128 and n <= st["prune_first_block"]
+        C = C.clone()
+        skm.skm_update(pc, a_c, C)
+        a_prev = a_w
+    # skm_fit on a second point set of the same shapes, in a workspace that
+    # holds the first set's state: the same result as in a fresh workspace
+    X2 = _points(n, d, seed=78)
+    X2d = X2.to(DEV).to(torch.bfloat16).view(torch.int16)
+    x2b = X2d.cpu().numpy().view(np.uint16)
+    C2 = torch.from_numpy(oracle.bf16_to_f32(x2b[synth.forgy_indices(n, k, seed=10).numpy()]).copy()).to(DEV)
+    p1 = skm.Points(skm.REPR_BF16, Xd, d, flags=skm.FLAG_PRUNE)
+    p2 = skm.Points(skm.REPR_BF16, X2d, d, flags=skm.FLAG_PRUNE)
+    wsf = skm.workspace(skm.OP_FIT, p1, k)
+    skm.skm_fit(p1, k, 4, C_init=C2.clone(), ws=wsf, want_objective=False)
+    Ca, aa, _, _, _ = skm.skm_fit(p2, k, 4, C_init=C2.clone(), ws=wsf, want_objective=False)
+    Cb, ab, _, _, _ = skm.skm_fit(p2, k, 4, C_init=C2.clone(), want_objective=False)
+    assert torch.equal(aa, ab) and torch.equal(Ca, Cb)
+
+
 @pytest.mark.parametrize("repr_name", ["bf16", "f32"])
 def test_warm_screen_bounds_across_lloyd_steps(skm, repr_name):
     """SKM_FLAG_WARM: each call starts every row's screen threshold from the
