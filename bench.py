@@ -408,18 +408,29 @@ def run_ours(args):
     # ---- inputs (per-rank shard), resident in HBM before timing -------------
     Yb, C, idx, proj = setup_head(dev, rank, world, dist, peaks)
     N, K = Yb.shape[0], C.shape[0]
-    # per-point norms built once; FLAG_WARM: the same points and assignment
-    # workspace every step, so each screen starts from the previous bounds
-    pts = skm.Points(skm.REPR_BF16, Yb, D_PCA, flags=0 if args.cold_screen else skm.FLAG_WARM).with_screen()
-    wsA = skm.workspace(skm.OP_ASSIGN, pts, K)
-    wsU = skm.workspace(skm.OP_UPDATE, pts, K)
+    warm = 0 if args.cold_screen else skm.FLAG_WARM
+    # the dense bf16 screen (per-point norms built once; FLAG_WARM: each screen
+    # starts from the previous call's bounds): the first step's seeds, and the
+    # comparison step (--dense)
+    pts_d = skm.Points(skm.REPR_BF16, Yb, D_PCA, flags=warm).with_screen()
+    wsD = skm.workspace(skm.OP_ASSIGN, pts_d, K)
+    # the step's assignment: exact dimension pruning (Section 3.1
+    # "SuperKMeans") with the first 128 dimensions on tensor cores, seeded with
+    # the previous step's assignment; FLAG_WARM: each row's bound carried over
+    pts_p = skm.Points(skm.REPR_BF16, Yb, D_PCA, flags=skm.FLAG_PRUNE | warm)
+    pts = pts_d if args.dense else pts_p
+    wsA = wsD if args.dense else skm.workspace(skm.OP_ASSIGN, pts_p, K)
+    wsU = skm.workspace(skm.OP_UPDATE, pts_d, K)
     a = torch.empty(N, dtype=torch.int32, device=dev)
+    skm.skm_assign(pts_d, C, K, want_dist=False, ws=wsD, out=a)  # seeds of the first step (setup)
+    a_seed = a.clone()
     cnt = torch.zeros(K, dtype=torch.int64, device=dev)
     part = torch.zeros(K, D_PCA, dtype=torch.float64, device=dev) if world > 1 else None
     C_step = C.clone()
+    prev = None if args.dense else a
 
     def step():
-        skm.skm_assign(pts, C_step, K, want_dist=False, ws=wsA, out=a)
+        skm.skm_assign(pts, C_step, K, prev_assign=prev, want_dist=False, ws=wsA, out=a)
         if part is None:
             skm.skm_update(pts, a, C_step, counts=cnt, ws=wsU)
         else:  # the one exchange: cluster sums and counts, all-reduced
@@ -438,29 +449,54 @@ def run_ours(args):
     # ---- per-kernel times (eager calls after the timed region) ----------------
     # assignment and update each timed inside eager steps (every assignment
     # after an update, as in the timed region)
-    t_assign, t_update = _split_ms([lambda: skm.skm_assign(pts, C_step, K, want_dist=False, ws=wsA, out=a),
+    t_assign, t_update = _split_ms([lambda: skm.skm_assign(pts, C_step, K, prev_assign=prev, want_dist=False,
+                                                           ws=wsA, out=a),
                                     lambda: skm.skm_update(pts, a, C_step, counts=cnt, ws=wsU)], 3, stream)
     long_region = ms > 1000.0
     bf16_peak = peaks["bf16_tflops_sustained"] if long_region else peaks["bf16_tflops"]
     flops = 2.0 * N * K * D_PCA
     upd_bytes = N * D_PCA * 2 + N * 4 * 3  # rows read once; assignments, sorted order, cluster ids
-    kernels = {
-        "assign_bf16_screen": {
-            "ms": t_assign, "bound": "tensor", "achieved": flops / (t_assign / 1e3) / 1e12, "peak": bf16_peak,
+    kernels = {}
+    if not args.dense:
+        st = skm.skm_assign_prune_stats(wsA, stream)  # the last split-timed call (a Lloyd step's)
+        F = st["prune_front_dims"]
+        fflops = 2.0 * N * K * F
+        kernels["assign_bf16_prune_front"] = {
+            "ms": t_assign, "bound": "tensor", "achieved": fflops / (t_assign / 1e3) / 1e12, "peak": bf16_peak,
             "unit": "TFLOP/s",
-            "algorithmic": f"2*N*k*d' = {flops:.3e} bf16 flop per launch (tensor-core screen; the call also "
-                           "prepares the centroids and rescores undecided rows in fp32)"},
+            "algorithmic": f"2*N*k*F = {fflops:.3e} bf16 flop per launch (F = {F} front dimensions on tensor cores, "
+                           "the measured executed work; the call also sorts the centroids, forms the rows' "
+                           "thresholds from their kept bounds and finishes the survivors on CUDA cores)",
+            "front_dims": F, "survivors_per_row": st["prune_first_block"] / N,
+            "rows_finished_cuda_cores": st["prune_rows_finished"], "rows_pruned_over_all_k": st["prune_rows_full"],
+            "cuda_core_block_sums": st["prune_blocks"], "complete_pairs": st["prune_complete"],
+            "dense_equivalent_tflops": flops / (t_assign / 1e3) / 1e12,
+            "note": "exact: the same assignments and distances as the CUDA-core prefix pruning, bit for bit"}
+        # the dense screen on the same centroids (warm from its own previous call)
+        a_d = torch.empty_like(a)
+        skm.skm_assign(pts_d, C_step, K, want_dist=False, ws=wsD, out=a_d)
+        t_dense = _event_ms(lambda: skm.skm_assign(pts_d, C_step, K, want_dist=False, ws=wsD, out=a_d), 3, stream)
+        kernels["assign_bf16_prune_front"]["agreement_with_dense_screen"] = float((a_d == a).float().mean())
+        del a_d
+    else:
+        t_dense = t_assign
+    kernels["assign_bf16_screen"] = {
+        "ms": t_dense, "bound": "tensor", "achieved": flops / (t_dense / 1e3) / 1e12, "peak": bf16_peak,
+        "unit": "TFLOP/s", "in_step": bool(args.dense),
+        "algorithmic": f"2*N*k*d' = {flops:.3e} bf16 flop per launch (dense tensor-core screen; the call also "
+                       "prepares the centroids and rescores undecided rows in fp32)"}
+    kernels.update({
         "update_bf16": {
             "ms": t_update, "bound": "hbm", "achieved": upd_bytes / (t_update / 1e3) / 1e9, "peak": peaks["hbm_gbs"],
             "unit": "GB/s", "algorithmic": f"N*d'*2 + 12*N = {upd_bytes:.3e} bytes per launch (bf16 rows read once, "
                                            "assignments, sorted order and cluster ids)"},
         "project_pca": proj,
-    }
+    })
 
     # ---- the pruned assignment of the same workload (exact, SKM_FLAG_PRUNE) on a row subset
     if not args.no_prune and world == 1:
         ns = min(N, 1_000_000)
-        pp = skm.Points(skm.REPR_BF16, Yb[:ns], D_PCA, flags=skm.FLAG_PRUNE)
+        pp = skm.Points(skm.REPR_BF16, Yb[:ns], D_PCA, flags=skm.FLAG_PRUNE | skm.FLAG_PRUNE_CUDA_CORES)
         ap = torch.empty(ns, dtype=torch.int32, device=dev)
         prev = a[:ns].clone()  # bound seeded with the previous assignment's centroid
         wsP = skm.workspace(skm.OP_ASSIGN, pp, K)
@@ -484,11 +520,12 @@ def run_ours(args):
     for kd in kernels.values():
         if "achieved" in kd:
             kd["frac"] = kd["achieved"] / kd["peak"]
-    kd = kernels["assign_bf16_screen"]
-    traffic = TRAFFIC_PER_POINT.get("assign_bf16_screen")
+    head_kernel = "assign_bf16_screen" if args.dense else "assign_bf16_prune_front"
+    kd = kernels[head_kernel]
+    traffic = TRAFFIC_PER_POINT.get(head_kernel)
     roofline = {"bound": kd["bound"], "achieved": round(kd["achieved"], 4), "peak": round(kd["peak"], 4),
                 "unit": kd["unit"], "frac": round(kd["frac"], 5),
-                "traffic": round(traffic * N) if traffic else None, "kernel": "assign_bf16_screen",
+                "traffic": round(traffic * N) if traffic else None, "kernel": head_kernel,
                 "peak_source": f"{peaks['source']} ({'sustained' if long_region else 'burst'} bf16)"}
 
     # ---- end to end through the C ABI with host buffers ----------------------
@@ -496,9 +533,13 @@ def run_ours(args):
     if not args.no_e2e:
         Y_host = torch.empty(N, D_PCA, dtype=torch.int16, pin_memory=True)
         Y_host.copy_(Yb)
+        # the Lloyd run continues from the device steps' centroids and
+        # assignments (the seeds of the first call; each call then leaves its
+        # assignments there)
         C_host = torch.empty(K, D_PCA, dtype=torch.float32, pin_memory=True)
-        C_host.copy_(C)
+        C_host.copy_(C_step)
         a_host = torch.empty(N, dtype=torch.int32, pin_memory=True)
+        a_host.copy_(a)
         holder = {}
 
         def exchange():
@@ -507,7 +548,8 @@ def run_ours(args):
             dist.all_reduce(s.counts)
 
         hstep = skm.LloydStepHost(skm.REPR_BF16, Y_host, D_PCA, K, chunks=E2E_CHUNKS, device=dev,
-                                  exchange=exchange if world > 1 else None, warm=not args.cold_screen)
+                                  exchange=exchange if world > 1 else None, warm=not args.cold_screen,
+                                  prune=not (args.dense or args.cold_screen))
         holder["step"] = hstep
         for _ in range(2):  # untimed warm-up (first-use costs of the range-sized calls)
             hstep(C_host, C_host, a_host)
@@ -536,16 +578,17 @@ def run_ours(args):
                "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "steps": e2e_steps,
                "ms_per_step": ems / e2e_steps, "h2d_probe_gbs": round(h2d_probe_gbs, 1),
                "h2d_effective_gbs": round(h2d / (ems / e2e_steps / 1e3) / 1e9, 1),
-               "path": f"skm_lloyd_step_host: pinned host bf16 points -> {E2E_CHUNKS} row ranges copied on a copy "
-                       "stream into three device range buffers while earlier ranges are assigned (each range's "
-                       "screen from the bounds its previous call left) and summed -> finalised centroids and "
-                       "assignments back in host memory on return (host wall clock per call)"}
+               "path": f"skm_lloyd_step_host: pinned host bf16 points (and, pruned, the previous assignments as "
+                       f"seeds) -> {E2E_CHUNKS} row ranges copied on a copy stream into three device range buffers "
+                       "while earlier ranges are assigned (each range from the bounds its previous call left) and "
+                       "summed -> finalised centroids and assignments back in host memory on return (host wall "
+                       "clock per call)"}
         del hstep, Y_host
 
     # ---- the other configurations (one GPU) -------------------------------------
     extra = None
     if world == 1 and not args.no_extra:
-        del wsA, wsU, pts
+        del wsA, wsU, pts, pts_d, pts_p, wsD
         torch.cuda.empty_cache()
         extra = run_extra_configs(args, dev, peaks, stream, local_rank)
 
@@ -562,10 +605,15 @@ def run_ours(args):
             "metric": METRIC, "value": value, "unit": "distances/s", "n_gpus": world, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": ms_step, "higher_is_better": True, "scaling": "weak",
             "vs_baseline": None,
-            "dtype": "bf16 points, fp32 centroids (bf16 tensor-core screen + fp32 rescore: the exact fp32 argmin)",
+            "dtype": ("bf16 points, fp32 centroids (bf16 tensor-core screen + fp32 rescore: the exact fp32 argmin)"
+                      if args.dense else
+                      "bf16 points, fp32 centroids (exact prefix pruning: bf16 tensor-core front over 128 dims "
+                      "with a rigorous bound, survivors finished in fp32 block sums: the exact fp32 argmin)"),
             "data": "synthetic (seeded GMM embeddings, generated on the GPU; PCA fitted on them)",
             "config": {"workload": WORKLOAD, "n": N, "D": 1024, "d": D_PCA, "k": K, "repr": "bf16 (PCA-256)",
-                       "step": "one Lloyd iteration (assign + update) over all points",
+                       "step": ("one Lloyd iteration (assign + update) over all points" + (
+                           "" if args.dense else "; assignment: exact dimension pruning seeded with the previous "
+                                                 "step's assignment, bounds carried between steps")),
                        "l2": "inputs larger than L2 (5.1 GB of bf16 points streamed every step)",
                        "timing": timing, "parallelism": f"dp{world}"},
             "roofline": roofline, "kernels": kernels, "configs": extra, "cpu_baseline": cpu, "e2e": e2e,
@@ -1052,7 +1100,9 @@ def main():
                          "update_lvq4|project|quantize_sq8|quantize_rbq1|quantize_lvq4")
     ap.add_argument("--n", type=int, default=200_000)
     ap.add_argument("--cold-screen", action="store_true",
-                    help="headline step without SKM_FLAG_WARM (every screen starts with no bound)")
+                    help="headline step without SKM_FLAG_WARM (every call starts with no carried bound)")
+    ap.add_argument("--dense", action="store_true",
+                    help="headline step with the dense bf16 screen instead of the pruned assignment")
     ap.add_argument("--e4m3-copy", action="store_true",
                     help="--case assign_rbq1 / assign_lvq4: read the points from their e4m3 copy instead of packed")
     ap.add_argument("--d", type=int, default=768)

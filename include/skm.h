@@ -116,7 +116,10 @@ enum {
      * ||c' - c||)^2 (1 + g) with g covering the fp32 rounding, and forms the
      * front's threshold from U' without reading the points.  Calls that want
      * distances use the exact seed distances instead. */
-    SKM_FLAG_WARM = 4
+    SKM_FLAG_WARM = 4,
+    /* With SKM_FLAG_PRUNE on BF16: no tensor-core front, the CUDA-core
+     * pruning kernels only (the same result; for comparisons). */
+    SKM_FLAG_PRUNE_CUDA_CORES = 8
 };
 
 /* Points being clustered.  Which fields are read depends on repr. */
@@ -645,7 +648,15 @@ typedef struct skm_step_host_config {
                                previous call left (SKM_FLAG_WARM); the
                                workspace then holds one assignment workspace
                                per range.  0: every call starts cold.        */
-    int32_t reserved[3];
+    int32_t prune;          /* BF16 with warm = 1: each range's assignment is
+                               the exact pruned one (SKM_FLAG_PRUNE, the
+                               tensor-core front), seeded with the previous
+                               call's assignments, which assign_host must
+                               hold on entry (the caller passes the array
+                               back unchanged; the first call's seeds decide
+                               only its work).  The range's seeds are copied
+                               in with its points.                           */
+    int32_t reserved[2];
 } skm_step_host_config;
 
 size_t skm_step_host_workspace_size(const skm_step_host_config *cfg, const skm_data *x);

@@ -24,7 +24,7 @@ __all__ = [
 ]
 
 REPR_F32, REPR_SQ8, REPR_RBQ1, REPR_BF16, REPR_LVQ4 = 0, 1, 2, 3, 4
-FLAG_PRUNE, FLAG_SYMMETRIC, FLAG_WARM = 1, 2, 4
+FLAG_PRUNE, FLAG_SYMMETRIC, FLAG_WARM, FLAG_PRUNE_CUDA_CORES = 1, 2, 4, 8
 DTYPE_F32, DTYPE_BF16 = 0, 1
 EMPTY_KEEP, EMPTY_SPLIT = 0, 1
 OP_ASSIGN, OP_UPDATE, OP_FIT, OP_QUANTIZE, OP_PCA, OP_ASSIGN_SEG = 0, 1, 2, 3, 4, 5
@@ -103,7 +103,8 @@ class StepHostConfig(ctypes.Structure):
 
     _fields_ = [("k", ctypes.c_int32), ("chunks", ctypes.c_int32), ("copy_stream", ctypes.c_void_p),
                 ("partial", ctypes.c_void_p), ("counts", ctypes.c_void_p), ("exchange", EXCHANGE_FN),
-                ("user", ctypes.c_void_p), ("warm", ctypes.c_int32), ("reserved", ctypes.c_int32 * 3)]
+                ("user", ctypes.c_void_p), ("warm", ctypes.c_int32), ("prune", ctypes.c_int32),
+                ("reserved", ctypes.c_int32 * 2)]
 
 
 def lib_path() -> str:
@@ -581,9 +582,13 @@ class LloydStepHost:
     enqueue its work on the step's stream and then reads/writes the tensors
     `self.partial` and `self.counts`.  warm=True: the host points do not
     change between calls, so each row range's screen starts from the bounds
-    its previous call left (one assignment workspace per range)."""
+    its previous call left (one assignment workspace per range).
+    prune=True (BF16, with warm): exact pruned assignments seeded with the
+    assignments in the assign_host array passed to the call (the previous
+    call's, passed back unchanged)."""
 
-    def __init__(self, repr_, X_host, d, k, chunks=16, device=None, copy_stream=None, exchange=None, warm=False):
+    def __init__(self, repr_, X_host, d, k, chunks=16, device=None, copy_stream=None, exchange=None, warm=False,
+                 prune=False):
         self.device = torch.device("cuda") if device is None else torch.device(device)
         self.repr, self.k, self.d = repr_, int(k), int(d)
         self.X_host = X_host
@@ -595,7 +600,8 @@ class LloydStepHost:
         self._user_exchange = exchange
         self._cb = EXCHANGE_FN(self._exchange) if exchange is not None else EXCHANGE_FN()
         self.cfg = StepHostConfig(self.k, int(chunks), ctypes.c_void_p(self.copy_stream.cuda_stream),
-                                  self.partial.data_ptr(), self.counts.data_ptr(), self._cb, None, int(bool(warm)))
+                                  self.partial.data_ptr(), self.counts.data_ptr(), self._cb, None, int(bool(warm)),
+                                  int(bool(prune)))
         nbytes = lib().skm_step_host_workspace_size(ctypes.byref(self.cfg), ctypes.byref(self.ref))
         if nbytes == 0:
             raise SkmError(1, lib().skm_last_error().decode())

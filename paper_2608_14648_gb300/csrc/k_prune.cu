@@ -14,6 +14,8 @@
 // non-negative, so dropping a centroid whose partial already exceeds beta
 // never drops the nearest one; `slack` covers the fp32 rounding of the sums,
 // so the result is the exact fp32 argmin whatever the seed.
+#include <climits>
+
 #include "skm_internal.cuh"
 
 namespace skm {
@@ -194,7 +196,7 @@ __global__ void __launch_bounds__(PRC_WARPS * 32) prune_rows_cta_kernel(
     const uint16_t *__restrict__ X, int d, const float *__restrict__ C, int k, const int32_t *__restrict__ seeds,
     const float2 *__restrict__ thr, int2 *__restrict__ wrow, const int32_t *__restrict__ rows,
     const int32_t *__restrict__ nrows, int32_t *__restrict__ assign, float *__restrict__ dist,
-    unsigned long long *__restrict__ counters) {
+    unsigned long long *__restrict__ counters, int max_rows) {
     __shared__ float sx[PR_MAX_D];
     __shared__ int qid[PRC_WARPS][2][PR_BATCH];
     __shared__ float qps[PRC_WARPS][2][PR_BATCH];
@@ -203,6 +205,7 @@ __global__ void __launch_bounds__(PRC_WARPS * 32) prune_rows_cta_kernel(
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const float slack = prune_slack(d);
     const int64_t nr = (int64_t)*nrows;
+    if (nr >= max_rows) return;  // the tiled kernel takes a list this long
     unsigned long long first_alive = 0, complete = 0, later = 0;
     for (int64_t ri = blockIdx.x; ri < nr; ri += gridDim.x) {
         const int64_t row = rows[ri];
@@ -409,11 +412,18 @@ __device__ __forceinline__ void survivor(unsigned M0, unsigned M1, int i, int &s
     owner = (i < n0 + __popc(M1)) ? (int)__fns(ms, 0, rank + 1) : 0;
 }
 
-template <typename TX>
+// rows (NULL: every row, one tile of TP_PTS points per CTA): a list of
+// *nrows rows walked tile by tile over the grid, whose seeds and seed
+// distances (or bounds) come from seeds / thr (the tensor-core front's rows
+// pruned over all k); with fewer than min_rows listed rows the kernel leaves
+// them to the one-CTA-per-row kernel.  wrow (optional): (distance bits,
+// centroid) of each row for the next call.
+template <typename TX, bool LIST>
 __global__ void __launch_bounds__(TP_WARPS * 32) prune_tiled_kernel(
     const TX *__restrict__ X, int64_t n, int d, const float *__restrict__ C, int k,
     const int32_t *__restrict__ prev, int32_t *__restrict__ assign, float *__restrict__ dist,
-    unsigned long long *__restrict__ counters) {
+    unsigned long long *__restrict__ counters, const int32_t *__restrict__ rows, const int32_t *__restrict__ nrows,
+    int min_rows, const int32_t *__restrict__ seeds, const float2 *__restrict__ thr, int2 *__restrict__ wrow) {
     extern __shared__ __align__(16) float tp_smem[];
     const int dp = ((d + 31) & ~31) + 4;  // padded centroid row (floats): a 16-byte multiple, banks shift by 4
     const int dx = (d + 31) & ~31;
@@ -424,23 +434,36 @@ __global__ void __launch_bounds__(TP_WARPS * 32) prune_tiled_kernel(
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int nb = (d + 31) >> 5;
     const float slack = 1.0f + 2.0f * (float)(d + 1) * 0x1p-24f;
-    const int64_t p0 = (int64_t)blockIdx.x * TP_PTS;
-    const int np = (int)min((int64_t)TP_PTS, n - p0);
+    const int64_t nr = LIST ? (int64_t)*nrows : n;
+    if (LIST && nr < min_rows) return;
     unsigned long long first_alive = 0, complete = 0, later = 0;
+    // a list: tiles over the grid; otherwise one tile per CTA
+    const int64_t pstep = LIST ? (int64_t)gridDim.x * TP_PTS : nr;
+    for (int64_t p0 = (int64_t)blockIdx.x * TP_PTS; p0 < nr; p0 += pstep) {
+    const int np = (int)min((int64_t)TP_PTS, nr - p0);
+    auto row_of = [&](int q) { return LIST ? (int64_t)rows[p0 + q] : p0 + q; };
+    __syncthreads();  // the previous tile's results are written
     for (int e = threadIdx.x; e < TP_PTS * dx; e += blockDim.x) {
         const int q = e / dx, i = e - q * dx;
-        xs[e] = (q < np && i < d) ? ldx<TX>(X + (p0 + q) * d + i) : 0.0f;
+        xs[e] = (q < np && i < d) ? ldx<TX>(X + row_of(q) * d + i) : 0.0f;
     }
     __syncthreads();
-    // each point's bound: its full distance to the seed centroid (block sums in order)
+    // each point's bound: its full distance to the seed centroid (block sums
+    // in order), or the listed row's seed distance (or bound) already formed
     for (int q = warp; q < np; q += TP_WARPS) {
-        int best = prev ? prev[p0 + q] : 0;
-        if (best < 0 || best >= k) best = 0;
+        const int64_t row = row_of(q);
         if (lane == 0) {
-            float beta = 0.0f;
-            for (int b = 0; b < nb; ++b) beta += block_partial(xs + q * dx, C + (int64_t)best * d, d, b);
-            s_beta[q] = beta;
-            s_best[q] = best;
+            if (LIST) {
+                s_beta[q] = thr[row].y;
+                s_best[q] = seeds[row];
+            } else {
+                int best = prev ? prev[row] : 0;
+                if (best < 0 || best >= k) best = 0;
+                float beta = 0.0f;
+                for (int b = 0; b < nb; ++b) beta += block_partial(xs + q * dx, C + (int64_t)best * d, d, b);
+                s_beta[q] = beta;
+                s_best[q] = best;
+            }
         }
     }
     for (int c0 = 0; c0 < k; c0 += TP_KC) {
@@ -528,9 +551,12 @@ __global__ void __launch_bounds__(TP_WARPS * 32) prune_tiled_kernel(
     }
     __syncthreads();
     for (int q = threadIdx.x; q < np; q += blockDim.x) {
-        assign[p0 + q] = s_best[q];
-        if (dist) dist[p0 + q] = s_beta[q];
+        const int64_t row = row_of(q);
+        assign[row] = s_best[q];
+        if (dist) dist[row] = s_beta[q];
+        if (LIST && wrow) wrow[row] = make_int2(__float_as_int(s_beta[q]), s_best[q]);
     }
+    }  // tiles
     if (counters) {
 #pragma unroll
         for (int o = 16; o > 0; o >>= 1) {
@@ -796,17 +822,19 @@ cudaError_t launch_prune_assign(const void *X, int x_is_bf16, int64_t n, int d, 
         const size_t smem = ((size_t)TP_KC * dp + (size_t)TP_PTS * dx + 2 * TP_PTS) * sizeof(float);
         const int64_t blocks = (n + TP_PTS - 1) / TP_PTS;
         if (x_is_bf16) {
-            cudaError_t e = cudaFuncSetAttribute(prune_tiled_kernel<uint16_t>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+            cudaError_t e = cudaFuncSetAttribute(prune_tiled_kernel<uint16_t, false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                                  (int)smem);
             if (e != cudaSuccess) return e;
-            prune_tiled_kernel<uint16_t><<<(unsigned)blocks, TP_WARPS * 32, smem, st>>>(
-                static_cast<const uint16_t *>(X), n, d, C, k, prev, assign, dist, counters);
+            prune_tiled_kernel<uint16_t, false><<<(unsigned)blocks, TP_WARPS * 32, smem, st>>>(
+                static_cast<const uint16_t *>(X), n, d, C, k, prev, assign, dist, counters, nullptr, nullptr, 0,
+                nullptr, nullptr, nullptr);
         } else {
-            cudaError_t e = cudaFuncSetAttribute(prune_tiled_kernel<float>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+            cudaError_t e = cudaFuncSetAttribute(prune_tiled_kernel<float, false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                                  (int)smem);
             if (e != cudaSuccess) return e;
-            prune_tiled_kernel<float><<<(unsigned)blocks, TP_WARPS * 32, smem, st>>>(
-                static_cast<const float *>(X), n, d, C, k, prev, assign, dist, counters);
+            prune_tiled_kernel<float, false><<<(unsigned)blocks, TP_WARPS * 32, smem, st>>>(
+                static_cast<const float *>(X), n, d, C, k, prev, assign, dist, counters, nullptr, nullptr, 0,
+                nullptr, nullptr, nullptr);
         }
         return launched();
     }
@@ -825,8 +853,21 @@ cudaError_t launch_prune_rows_cta(const uint16_t *X, int d, const float *C, int 
                                   const int32_t *rows, const int32_t *nrows, int32_t *assign,
                                   float *dist, unsigned long long *counters, cudaStream_t st) {
     if (d > PR_MAX_D) return cudaErrorInvalidValue;
+    // a long list (d <= 256): the tiled kernel (centroid chunks staged once
+    // per TP_PTS rows); a short one: one CTA per row (more rows in flight)
+    const bool tiled = d <= TP_MAX_D_F32 && (reinterpret_cast<uintptr_t>(C) & 15) == 0;
+    constexpr int LONG_LIST = 8192;
     prune_rows_cta_kernel<<<152 * 4, PRC_WARPS * 32, 0, st>>>(X, d, C, k, r.seed, r.thr, r.wrow, rows, nrows, assign,
-                                                              dist, counters);
+                                                              dist, counters, tiled ? LONG_LIST : INT_MAX);
+    cudaError_t e = launched();
+    if (e != cudaSuccess || !tiled) return e;
+    const int dx = (d + 31) & ~31, dp = dx + 4;
+    const size_t smem = ((size_t)TP_KC * dp + (size_t)TP_PTS * dx + 2 * TP_PTS) * sizeof(float);
+    e = cudaFuncSetAttribute(prune_tiled_kernel<uint16_t, true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             (int)smem);
+    if (e != cudaSuccess) return e;
+    prune_tiled_kernel<uint16_t, true><<<152, TP_WARPS * 32, smem, st>>>(X, 0, d, C, k, nullptr, assign, dist, counters,
+                                                                    rows, nrows, LONG_LIST, r.seed, r.thr, r.wrow);
     return launched();
 }
 

@@ -164,7 +164,8 @@ static void plan_assign(const skm_data *x, int k, Carver &cv, AssignBufs &b) {
         }
         tc_plan(-1, n, d, k, x->x, x->screen, false, cv, b.tc);  // statistics only
         // bf16 points: the tensor-core front, taken when a seed assignment is given
-        if (tc_pfront_ok(x->repr, d, x->x)) tc_plan_pfront(n, d, k, (x->flags & SKM_FLAG_WARM) != 0, cv, b.tc);
+        if (tc_pfront_ok(x->repr, d, x->x) && !(x->flags & SKM_FLAG_PRUNE_CUDA_CORES))
+            tc_plan_pfront(n, d, k, (x->flags & SKM_FLAG_WARM) != 0, cv, b.tc);
         return;
     }
     switch (x->repr) {

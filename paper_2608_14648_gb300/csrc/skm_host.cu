@@ -44,6 +44,8 @@ int host_check(const skm_step_host_config *cfg, const skm_data *x) {
     if (cfg->chunks < 1 || cfg->chunks > MAX_CHUNKS)
         return set_error(SKM_ERR_INVALID_ARG, "chunks = %d outside [1, %d]", cfg->chunks, MAX_CHUNKS);
     if (x->screen) return set_error(SKM_ERR_INVALID_ARG, "skm_lloyd_step_host: x->screen must be NULL");
+    if (cfg->prune && (!cfg->warm || x->repr != SKM_REPR_BF16))
+        return set_error(SKM_ERR_UNSUPPORTED, "skm_lloyd_step_host: prune needs warm and BF16 points");
     return SKM_OK;
 }
 
@@ -93,6 +95,7 @@ void plan_host(const skm_step_host_config *cfg, const skm_data *x, Carver &cv, H
     // every range: the compute stream runs them one after another)
     skm_data probe = view_of(x, reinterpret_cast<const void *>(256), rc);
     if (host_warm(cfg, x)) probe.flags |= SKM_FLAG_WARM;
+    if (cfg->prune) probe.flags |= SKM_FLAG_PRUNE;
     b.ws_a_bytes = skm_workspace_size(0, &probe, k);
     probe.flags = 0;
     b.ws_u_bytes = skm_workspace_size(1, &probe, k);
@@ -185,6 +188,9 @@ extern "C" int skm_lloyd_step_host(const skm_step_host_config *cfg, const skm_da
             if (rows <= 0) break;
             if (i >= nr) SKM_CUDA_TRY(cudaStreamWaitEvent(cp, freed[s], 0));
             SKM_CUDA_TRY(cudaMemcpyAsync(b.ring[s], xh + r0 * rb, (size_t)(rows * rb), cudaMemcpyHostToDevice, cp));
+            if (cfg->prune)  // the range's seeds: the previous call's assignments
+                SKM_CUDA_TRY(cudaMemcpyAsync(b.assign[s], assign_host + r0, sizeof(int32_t) * (size_t)rows,
+                                             cudaMemcpyHostToDevice, cp));
             SKM_CUDA_TRY(cudaEventRecord(landed[s], cp));
             SKM_CUDA_TRY(cudaStreamWaitEvent(st, landed[s], 0));
             skm_data v = view_of(x, b.ring[s], rows);
@@ -193,8 +199,9 @@ extern "C" int skm_lloyd_step_host(const skm_step_host_config *cfg, const skm_da
                 v.flags |= SKM_FLAG_WARM;
                 wsa = b.ws_a + (size_t)i * b.ws_a_stride;
             }
-            SKM_TRY(skm_assign(&v, b.C, k, nullptr, b.assign[s], objective_host ? b.dist[s] : nullptr, wsa,
-                               b.ws_a_bytes, st));
+            if (cfg->prune) v.flags |= SKM_FLAG_PRUNE;
+            SKM_TRY(skm_assign(&v, b.C, k, cfg->prune ? b.assign[s] : nullptr, b.assign[s],
+                               objective_host ? b.dist[s] : nullptr, wsa, b.ws_a_bytes, st));
             v.flags = 0;
             SKM_TRY(skm_update(&v, b.assign[s], k, nullptr, counts, partial, b.ws_u, b.ws_u_bytes, st));
             if (objective_host) {

@@ -188,6 +188,22 @@ def test_step_host_arguments_are_rejected_before_any_work(skm):
     x8 = skm.Data(1, 16, 100, X.ctypes.data, None, None, None, None, 0, 0)
     assert L.skm_step_host_workspace_size(ctypes.byref(warm), ctypes.byref(x8)) == \
         L.skm_step_host_workspace_size(ctypes.byref(cfg()), ctypes.byref(x8))
+    # prune: BF16 with warm only; the ranges' workspaces then hold survivor lists
+    Xb = np.zeros((1000, 256), np.uint16)
+    xb = skm.Data(skm.REPR_BF16, 256, 1000, Xb.ctypes.data, None, None, None, None, 0, 0)
+    pr = cfg()
+    pr.warm, pr.prune = 1, 1
+    wb = cfg()
+    wb.warm = 1
+    assert L.skm_step_host_workspace_size(ctypes.byref(pr), ctypes.byref(xb)) >= \
+        L.skm_step_host_workspace_size(ctypes.byref(wb), ctypes.byref(xb)) + 1000 * 256
+    cold_prune = cfg()
+    cold_prune.prune = 1
+    for c, xx in ((cold_prune, xb), (pr, x)):  # without warm; F32 points
+        assert L.skm_step_host_workspace_size(ctypes.byref(c), ctypes.byref(xx)) == 0
+        assert L.skm_lloyd_step_host(ctypes.byref(c), ctypes.byref(xx), FAKE, FAKE, FAKE, None, None, FAKE,
+                                     1 << 30, None) == 2
+        assert b"prune" in L.skm_last_error()
     for c, code, what in [(cfg(k=101), 1, b"k = 101"), (cfg(k=0), 1, b"k = 0"), (cfg(chunks=0), 1, b"chunks"),
                           (cfg(chunks=257), 1, b"chunks")]:
         assert L.skm_step_host_workspace_size(ctypes.byref(c), ctypes.byref(x)) == 0

@@ -142,3 +142,35 @@ def test_step_host_warm_ranges_match_cold(skm, kind, chunks):
         assert agree >= 0.9999, f"iteration {it}: agreement {agree}"
         if agree == 1.0:
             _close_l2(Cw, Cc)
+
+
+def test_step_host_pruned_ranges_match_device_pruning(skm):
+    """prune=1 (BF16, warm): each range's assignment is the exact pruned one
+    (tensor-core front seeded with the assignments passed in assign_host,
+    bounds kept per range); over Lloyd iterations it equals the device-side
+    pruned assignment bit for bit, and the centroids follow."""
+    n, d, k, chunks = 30000, 256, 300, 4
+    repr_, Xh, C0 = _inputs(skm, "bf16", n, d, k, seed=43)
+    Xp = Xh.pin_memory()
+    Xd = Xh.cuda()
+    pc = skm.Points(skm.REPR_BF16, Xd, d, flags=skm.FLAG_PRUNE)
+    dense = skm.Points(skm.REPR_BF16, Xd, d)
+    hstep = skm.LloydStepHost(repr_, Xp, d, k, chunks=chunks, warm=True, prune=True)
+    warm_only = skm.LloydStepHost(repr_, Xp, d, k, chunks=chunks, warm=True)
+    assert hstep.ws.numel() > warm_only.ws.numel()
+    a0, _ = skm.skm_assign(dense, C0.cuda())  # the first call's seeds
+    a_host = a0.cpu().pin_memory()
+    C = C0.clone().pin_memory()
+    for it in range(4):
+        a_ref, _ = skm.skm_assign(pc, C.cuda())
+        part = torch.zeros(k, d, dtype=torch.float64, device="cuda")
+        cnt = torch.zeros(k, dtype=torch.int64, device="cuda")
+        skm.skm_update(pc, a_ref, None, counts=cnt, partial=part)
+        C_ref = C.cuda().clone()
+        skm.skm_update_finalize(pc, part, cnt, C_ref)
+        torch.cuda.synchronize()
+        C_out = torch.empty_like(C).pin_memory()
+        hstep(C, C_out, a_host)
+        assert torch.equal(a_host, a_ref.cpu()), f"iteration {it}"
+        _close_l2(C_out, C_ref.cpu())
+        C = C_out
