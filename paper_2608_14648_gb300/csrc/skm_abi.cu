@@ -226,9 +226,35 @@ static void plan_update(const skm_data *x, int k, Carver &cv, UpdateBufs &b) {
     b.wsplit = cv.take<int64_t>(k);
 }
 
+// skm_fit with SKM_FLAG_PRUNE on points the tensor-core front takes: the
+// dense screen (a2) runs the iterations in which prefix pruning cannot pay
+// (the first, and while more than one in FIT_MOVED_DIV of the rows change
+// cluster), the pruned assignment (a) the later ones; a pruned iteration
+// that keeps more than FIT_MAX_SURVIVORS centroids a row sends the next one
+// back to the screen.  Both give the exact fp32 nearest centroid (they may
+// break a tie within fp32 rounding differently).
+constexpr int64_t FIT_MOVED_DIV = 100;
+constexpr double FIT_MAX_SURVIVORS = 8.0;
+static bool fit_front(const skm_data *x) {
+    return use_prune(x) && tc_pfront_ok(x->repr, x->d, x->x) && !(x->flags & SKM_FLAG_PRUNE_CUDA_CORES);
+}
+
+__global__ void count_moved_kernel(const int32_t *__restrict__ a, const int32_t *__restrict__ b, int64_t n,
+                                   unsigned long long *__restrict__ out) {
+    unsigned long long c = 0;
+    for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < n; i += (int64_t)gridDim.x * blockDim.x)
+        c += a[i] != b[i];
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) c += __shfl_xor_sync(0xffffffffu, c, o);
+    if ((threadIdx.x & 31) == 0 && c) atomicAdd(out, c);
+}
+
 struct FitBufs {
     uint8_t *screen = nullptr;  // built once per fit when the caller gave none
     AssignBufs a;
+    AssignBufs a2;                           // fit_front: the dense screen's
+    int32_t *aprev = nullptr;                // fit_front: the previous iteration's assignment
+    unsigned long long *moved = nullptr;     // fit_front: rows that changed cluster
     UpdateBufs u;
     float *dist = nullptr;
     double *partials = nullptr, *sum = nullptr;
@@ -253,6 +279,13 @@ static void plan_fit(const skm_data *x, int k, Carver &cv, FitBufs &b) {
         }
     }
     plan_assign(&xs, k, cv, b.a);
+    if (fit_front(x)) {
+        skm_data xd = xs;
+        xd.flags &= ~SKM_FLAG_PRUNE;
+        plan_assign(&xd, k, cv, b.a2);
+        b.aprev = cv.take<int32_t>(x->n);
+        b.moved = cv.take<unsigned long long>(1);
+    }
     plan_update(x, k, cv, b.u);
     b.dist = cv.take<float>(x->n);
     b.partials = cv.take<double>(RED_BLOCKS);
@@ -1162,8 +1195,14 @@ int skm_fit(const skm_fit_config *cfg, const skm_data *x, const void *C_init,
     // the iterations' screens start from the bounds the previous one left; the
     // first starts cold whatever state the workspace held (other points)
     if (x->repr == SKM_REPR_F32 || x->repr == SKM_REPR_BF16) xd.flags |= SKM_FLAG_WARM;
-    if (b.a.tc.warm_hdr) SKM_CUDA_TRY(cudaMemsetAsync(b.a.tc.warm_hdr, 0, 4 * sizeof(int64_t), st));
-    if (b.a.tc.pf_whdr) SKM_CUDA_TRY(cudaMemsetAsync(b.a.tc.pf_whdr, 0, 4 * sizeof(int64_t), st));
+    for (AssignBufs *ab : {&b.a, &b.a2}) {
+        if (ab->tc.warm_hdr) SKM_CUDA_TRY(cudaMemsetAsync(ab->tc.warm_hdr, 0, 4 * sizeof(int64_t), st));
+        if (ab->tc.pf_whdr) SKM_CUDA_TRY(cudaMemsetAsync(ab->tc.pf_whdr, 0, 4 * sizeof(int64_t), st));
+    }
+    const bool adaptive = fit_front(x);
+    skm_data xdense = xd;
+    xdense.flags &= ~SKM_FLAG_PRUNE;
+    if (adaptive) SKM_TRY(tc_init_stats(b.a2.tc, st));
     SKM_TRY(tc_init_stats(b.a.tc, st));
     SKM_CUDA_TRY(cudaMemsetAsync(b.a.prune, 0, PRUNE_CTRS * sizeof(unsigned long long), st));
     int e = 0;
@@ -1217,10 +1256,36 @@ int skm_fit(const skm_fit_config *cfg, const skm_data *x, const void *C_init,
     float *dist = dist_out ? dist_out : b.dist;
     const int nblk = (int)std::min<int64_t>(RED_BLOCKS, n);
     int32_t *assign = assign_out;
+    bool pruning = false;                 // adaptive: the pruned assignment is in use
+    unsigned long long surv_seen = 0;     // adaptive: front survivors counted so far
     for (int it = 0; it <= cfg->iters; ++it) {
         const bool want_obj = objective_host != nullptr;
-        SKM_TRY(do_assign(&xd, C_out, k, it > 0 ? assign : nullptr, assign,
-                          (want_obj || it == cfg->iters) ? dist : nullptr, b.a, st));
+        float *dist_it = (want_obj || it == cfg->iters) ? dist : nullptr;
+        if (adaptive && !pruning) {
+            if (it > 0)
+                SKM_CUDA_TRY(cudaMemcpyAsync(b.aprev, assign, sizeof(int32_t) * (size_t)n, cudaMemcpyDeviceToDevice,
+                                             st));
+            SKM_TRY(do_assign(&xdense, C_out, k, nullptr, assign, dist_it, b.a2, st));
+            if (it > 0 && it < cfg->iters) {  // settled enough for pruning to pay?
+                unsigned long long moved = 0;
+                SKM_CUDA_TRY(cudaMemsetAsync(b.moved, 0, sizeof(moved), st));
+                count_moved_kernel<<<(int)std::min<int64_t>(152 * 8, (n + 255) / 256), 256, 0, st>>>(assign, b.aprev,
+                                                                                             n, b.moved);
+                SKM_CUDA_TRY(launched());
+                SKM_CUDA_TRY(cudaMemcpyAsync(&moved, b.moved, sizeof(moved), cudaMemcpyDeviceToHost, st));
+                SKM_CUDA_TRY(cudaStreamSynchronize(st));
+                pruning = (int64_t)moved * FIT_MOVED_DIV <= n;
+            }
+        } else {
+            SKM_TRY(do_assign(&xd, C_out, k, it > 0 ? assign : nullptr, assign, dist_it, b.a, st));
+            if (adaptive && it < cfg->iters) {  // still pruning well?
+                unsigned long long surv = 0;
+                SKM_CUDA_TRY(cudaMemcpyAsync(&surv, b.a.prune, sizeof(surv), cudaMemcpyDeviceToHost, st));
+                SKM_CUDA_TRY(cudaStreamSynchronize(st));
+                pruning = (double)(surv - surv_seen) <= FIT_MAX_SURVIVORS * (double)n;
+                surv_seen = surv;
+            }
+        }
         if (want_obj) {
             SKM_CUDA_TRY(launch_sum_float_to_double(dist, n, b.partials, nblk, st));
             SKM_CUDA_TRY(launch_sum_double(b.partials, nblk, b.sum, st));
@@ -1245,6 +1310,13 @@ int skm_fit(const skm_fit_config *cfg, const skm_data *x, const void *C_init,
     skm_stats local;
     memset(&local, 0, sizeof(local));
     SKM_TRY(tc_read_stats(b.a.tc, &local, st));
+    if (adaptive) {  // the dense screen's iterations
+        skm_stats l2;
+        memset(&l2, 0, sizeof(l2));
+        SKM_TRY(tc_read_stats(b.a2.tc, &l2, st));
+        local.rescored_rows += l2.rescored_rows;
+        local.fallback_rows += l2.fallback_rows;
+    }
     int32_t uflag = 0;
     SKM_CUDA_TRY(cudaMemcpy(&uflag, b.u.flag, sizeof(uflag), cudaMemcpyDeviceToHost));
     if (uflag) return set_error(SKM_ERR_TIMEOUT, "an update pipeline wait exceeded its limit");
