@@ -188,6 +188,17 @@ typedef struct skm_stats {
 } skm_stats;
 
 const char *skm_last_error(void);
+
+/* Kernel timer, for profiling callers (the paper has no counterpart).  With
+ * skm_kernel_timer(1), CUDA events are recorded on the launch stream right
+ * before and after every tensor-core kernel launch (assignment, projection);
+ * skm_kernel_timer_ms waits for the later event and returns the time between
+ * the two, i.e. the last such launch's duration.  0 disables it (no events
+ * recorded).  Not for calls captured into a CUDA graph.  Errors:
+ * SKM_ERR_CUDA (event creation), SKM_ERR_INVALID_ARG (NULL ms, or never
+ * enabled). */
+int skm_kernel_timer(int on);
+int skm_kernel_timer_ms(float *ms);
 int skm_version(void); /* major*10000 + minor*100 + patch */
 
 /* Fault injection, for tests of the error paths (the paper has no

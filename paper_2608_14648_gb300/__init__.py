@@ -39,7 +39,7 @@ EXPORTED_SYMBOLS = [
     "skm_screen_prep", "skm_project", "skm_project_hadamard", "skm_unproject", "skm_copy_from_host",
     "skm_make_rotation",
     "skm_pca_fit", "skm_quantize", "skm_rbq1_exponent", "skm_lvq4_exponent", "skm_assign",
-    "skm_assign_prune_stats", "skm_assign_rbq1_noalloc",
+    "skm_assign_prune_stats", "skm_assign_rbq1_noalloc", "skm_kernel_timer", "skm_kernel_timer_ms",
     "skm_assign_segmented",
     "skm_update",
     "skm_merge_partials", "skm_update_finalize", "skm_fit", "skm_split_empty", "skm_hier_workspace_size",
@@ -138,6 +138,8 @@ def lib():
             "skm_lvq4_exponent": ([vp, i64, vp, vp, sz, vp], i32),
             "skm_assign": ([vp, vp, i32, vp, vp, vp, vp, sz, vp], i32),
             "skm_assign_prune_stats": ([vp, sz, vp, vp], i32),
+            "skm_kernel_timer": ([i32], i32),
+            "skm_kernel_timer_ms": ([vp], i32),
             "skm_assign_rbq1_noalloc": ([vp, vp, i32, vp, vp, vp], i32),
             "skm_assign_segmented": ([vp, vp, i32, vp, vp, i32, vp, vp, vp, sz, vp], i32),
             "skm_update": ([vp, vp, i32, vp, vp, vp, vp, sz, vp], i32),
@@ -423,6 +425,18 @@ def skm_assign(pts: Points, C, k=None, prev_assign=None, want_dist=True, ws=None
     _check(lib().skm_assign(ctypes.byref(pts.ref), _ptr(C), int(k), _ptr(prev_assign), _ptr(assign), _ptr(dist),
                             _ptr(ws), ws.numel(), _stream(stream)))
     return assign, dist
+
+
+def skm_kernel_timer(on):
+    """Enables (True) or disables the events around each tensor-core kernel launch."""
+    _check(lib().skm_kernel_timer(int(bool(on))))
+
+
+def skm_kernel_timer_ms():
+    """Duration (ms) of the last tensor-core kernel launch timed (waits for it)."""
+    ms = ctypes.c_float(0.0)
+    _check(lib().skm_kernel_timer_ms(ctypes.byref(ms)))
+    return float(ms.value)
 
 
 def skm_assign_prune_stats(ws, stream=None):

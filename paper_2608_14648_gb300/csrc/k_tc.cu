@@ -2147,7 +2147,9 @@ int launch_tc_kind(const void *xs, int64_t n, int dp, int d, const void *cs, int
     p.nct = (int)cdiv(k, BN);
     p.nkc = (int)cdiv(d, 128 / eb);
     p.inject_wait_ns = fault_take(SKM_FAULT_WAIT) ? 1000000ull : 0ull;  // 1 ms
+    tc_timer_mark(st, 0);
     kern<<<grid, tc_threads<NH, PK>(), SMEM, st>>>(ma, mb, p);
+    tc_timer_mark(st, 1);
     SKM_CUDA_TRY(launched());
     return SKM_OK;
 }

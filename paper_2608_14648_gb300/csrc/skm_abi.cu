@@ -41,6 +41,17 @@ bool fault_take(int kind) {
     return false;
 }
 
+// ---- timer of the tensor-core kernel launches (profiling callers)
+static std::mutex g_timer_mu;
+static std::atomic<int> g_timer_on{0};
+static cudaEvent_t g_timer_ev[2] = {nullptr, nullptr};
+
+void tc_timer_mark(cudaStream_t st, int which) {
+    if (!g_timer_on.load(std::memory_order_relaxed)) return;
+    std::lock_guard<std::mutex> lock(g_timer_mu);
+    if (g_timer_ev[which]) cudaEventRecord(g_timer_ev[which], st);
+}
+
 cudaError_t launched(int count) {
     g_launches.fetch_add((unsigned long long)count, std::memory_order_relaxed);
     const cudaError_t e = cudaGetLastError();
@@ -472,6 +483,28 @@ int skm_fault_armed(int kind) {
 int skm_version(void) { return 100; }
 
 uint64_t skm_kernel_launches(void) { return (uint64_t)g_launches.load(std::memory_order_relaxed); }
+
+int skm_kernel_timer(int on) {
+    std::lock_guard<std::mutex> lock(g_timer_mu);
+    if (on) {
+        for (auto &e : g_timer_ev)
+            if (!e && cudaEventCreate(&e) != cudaSuccess) {
+                e = nullptr;
+                return set_error(SKM_ERR_CUDA, "cudaEventCreate failed");
+            }
+    }
+    g_timer_on.store(on ? 1 : 0);
+    return SKM_OK;
+}
+
+int skm_kernel_timer_ms(float *ms) {
+    if (!ms) return set_error(SKM_ERR_INVALID_ARG, "ms is NULL");
+    std::lock_guard<std::mutex> lock(g_timer_mu);
+    if (!g_timer_ev[0] || !g_timer_ev[1]) return set_error(SKM_ERR_INVALID_ARG, "the timer was never enabled");
+    SKM_CUDA_TRY(cudaEventSynchronize(g_timer_ev[1]));
+    SKM_CUDA_TRY(cudaEventElapsedTime(ms, g_timer_ev[0], g_timer_ev[1]));
+    return SKM_OK;
+}
 
 size_t skm_workspace_size(int op, const skm_data *x, int k) {
     Carver cv(nullptr, 0);

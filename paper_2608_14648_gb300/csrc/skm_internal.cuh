@@ -36,6 +36,9 @@ cudaError_t launched(int count = 1);
 // True (and one armed occurrence used up) when an SKM_FAULT_* of this kind
 // is armed (skm_inject_fault or the SKM_FAULT environment variable).
 bool fault_take(int kind);
+// the kernel timer's events around a tensor-core kernel launch (which = 0
+// before, 1 after; nothing unless skm_kernel_timer enabled it)
+void tc_timer_mark(cudaStream_t st, int which);
 
 // ---- workspace carving ------------------------------------------------------
 // Sub-buffers are carved from the caller's workspace at 256-byte boundaries.

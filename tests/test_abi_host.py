@@ -158,6 +158,12 @@ def test_symmetric_flag_is_validated(skm):
     assert L.skm_workspace_size(0, ctypes.byref(r), 4) > 0
 
 
+def test_kernel_timer_arguments(skm):
+    L = skm.lib()
+    assert L.skm_kernel_timer_ms(None) == 1  # NULL output: rejected before any CUDA call
+    assert L.skm_kernel_timer(0) == 0  # disabling needs no device
+
+
 def test_copy_from_host_arguments(skm):
     L = skm.lib()
     FAKE = ctypes.c_void_p(0x1000)

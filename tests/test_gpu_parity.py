@@ -1467,3 +1467,26 @@ def test_fit_rbq1_segment_pruning_trajectory_bitexact(skm):
     np.testing.assert_array_equal(a.cpu().numpy(), ao)
     np.testing.assert_array_equal(C.cpu().numpy(), Co)
     assert 0 < st["prune_complete"] < st["prune_first_block"] < (iters + 1) * n * k
+
+
+def test_kernel_timer_times_the_tensor_core_launch(skm):
+    """skm_kernel_timer: events around each tensor-core kernel launch; the
+    last launch's duration is positive and below the whole call's."""
+    n, d, k = 50000, 256, 1000
+    X = _points(n, d, seed=91)
+    Xd = X.to(DEV).to(torch.bfloat16).view(torch.int16)
+    C = (Xd[synth.forgy_indices(n, k, seed=3).to(DEV)].to(torch.int32) << 16).view(torch.float32).contiguous()
+    pts = skm.Points(skm.REPR_BF16, Xd, d).with_screen()
+    ws = skm.workspace(skm.OP_ASSIGN, pts, k)
+    skm.skm_assign(pts, C, ws=ws)
+    skm.skm_kernel_timer(True)
+    try:
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record()
+        skm.skm_assign(pts, C, ws=ws)
+        e1.record()
+        ms = skm.skm_kernel_timer_ms()
+        torch.cuda.synchronize()
+        assert 0.0 < ms <= e0.elapsed_time(e1)
+    finally:
+        skm.skm_kernel_timer(False)
