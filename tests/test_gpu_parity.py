@@ -568,7 +568,7 @@ def test_prune_assign_vs_oracle_and_seed_independent(skm, repr_name, n, d, k):
 
 
 @pytest.mark.parametrize("n,d,k", [(3000, 256, 1000), (1000, 512, 300), (700, 1024, 257), (5000, 256, 13),
-                                   (130, 256, 600), (20000, 256, 1000)])
+                                   (130, 256, 600), (20000, 256, 1000), (1500, 264, 300), (900, 1000, 200)])
 def test_prune_front_tensor_cores_bitexact(skm, n, d, k):
     """bf16 points with a seed assignment: the first 128 dimensions of every
     pair screened on tensor cores, survivors finished on CUDA cores (Section
