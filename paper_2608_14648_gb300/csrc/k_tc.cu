@@ -1182,15 +1182,28 @@ __global__ void __launch_bounds__(tc_threads<NH, PK>(), 1)
                     // Records past k have ||c_F||^2 = +inf.  The slices take
                     // alternate chunks (neighbouring positions, which similar
                     // survivors tend to share, go to different sub-lists).
+                    // The warp releases the accumulator right after its last TMEM
+                    // load, so the MMA can refill it while that chunk is evaluated.
                     const float *cmins = reinterpret_cast<const float *>(rbuf + 1024);
                     const uint32_t tbase = tmem + ((uint32_t)(q * 32) << 16) + b * BN;
+                    int nvc = 0;  // this slice's chunks inside [0, k) (warp-uniform)
+                    while (nvc < SW / 32 && ct * BN + (NHG * nvc + slice) * 32 < p.k) ++nvc;
+                    if (nvc == 0) {
+                        tc_fence_before();
+                        __syncwarp();
+                        if (lane == 0) mbar_arrive(tempty_bar(b));
+                    }
 #pragma unroll 1
-                    for (int c = 0; c < SW / 32; ++c) {
+                    for (int c = 0; c < nvc; ++c) {
                         const int cc = (NHG * c + slice) * 32;  // column offset within the tile
                         const int j0 = ct * BN + cc;
-                        if (j0 >= p.k) break;  // warp-uniform
                         uint32_t v[32];
                         tmem_ld32(tbase + cc, v);
+                        if (c == nvc - 1) {  // the warp's loads are complete (each thread waited)
+                            tc_fence_before();
+                            __syncwarp();
+                            if (lane == 0) mbar_arrive(tempty_bar(b));
+                        }
                         auto f = [&](int i) { return __uint_as_float(v[i]); };
                         float m[11];
 #pragma unroll
@@ -1324,10 +1337,13 @@ __global__ void __launch_bounds__(tc_threads<NH, PK>(), 1)
                     }
                 }
                 // the warp's TMEM loads are complete (each thread waited on
-                // them); one arrival for the warp releases its share
-                tc_fence_before();
-                __syncwarp();
-                if (lane == 0) mbar_arrive(tempty_bar(b));
+                // them); one arrival for the warp releases its share (PFRONT:
+                // released after its last load already)
+                if (MODE != MODE_PFRONT) {
+                    tc_fence_before();
+                    __syncwarp();
+                    if (lane == 0) mbar_arrive(tempty_bar(b));
+                }
             }
             // merge the column slices of each row: slices 1.. publish, slice 0 finishes
             // (single buffer: a publisher rewrites its slot only at the end of
