@@ -64,6 +64,61 @@ __device__ __forceinline__ float block_partial(const float *sx, const float *c, 
     return s;
 }
 
+// Coalesced gather of 32 (centroid, block) pairs, one per lane: the warp
+// copies pair p's block (row j_p of C, dims [32 b_p, min(32 b_p + 32, d)))
+// to stg + p * STG_LD with 16-byte cp.async copies (no registers held, eight
+// in flight a lane), eight lanes per 128-byte block, so one instruction
+// touches four lines instead of one line per lane; each lane then reads its
+// own block from shared memory (rows 144 bytes apart: the eight lanes of a
+// 16-byte access phase hit distinct banks).  Needs d % 4 == 0, C 16-byte
+// aligned and k d <= 2^26.  Lanes with `valid` false stage nothing.
+constexpr int STG_LD = 36;
+__device__ __forceinline__ void stage_blocks(float *stg, const float *__restrict__ C, int d, int j, int b,
+                                             bool valid) {
+    const int lane = threadIdx.x & 31, q = lane & 7;
+    // (element offset of the block) * 16 + its length in float4s
+    const int key = valid ? (j * d + 32 * b) * 16 + (min(32, d - 32 * b) >> 2) : 0;
+    const uint32_t s0 = (uint32_t)__cvta_generic_to_shared(stg) + 16u * q;
+    __syncwarp();  // every lane has read the previous pairs
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+        const int p = 4 * i + (lane >> 3);
+        const int kp = __shfl_sync(0xffffffffu, key, p);
+        if (q < (kp & 15))
+            asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(s0 + (uint32_t)(p * STG_LD * 4)),
+                         "l"(C + (kp >> 4) + 4 * q)
+                         : "memory");
+    }
+    asm volatile("cp.async.commit_group;\n\tcp.async.wait_group 0;" ::: "memory");
+    __syncwarp();
+}
+// block_partial with the centroid block from shared memory (stage_blocks):
+// the same terms in the same order, so the same value
+__device__ __forceinline__ float block_partial_staged(const float *sx, const float *cb, int d, int b) {
+    float s = 0.0f;
+    const int i0 = 32 * b;
+    if (i0 + 32 <= d) {
+#pragma unroll
+        for (int q = 0; q < 8; ++q) {
+            const float4 cv = reinterpret_cast<const float4 *>(cb)[q];
+            float t = __fsub_rn(sx[i0 + 4 * q], cv.x);
+            s = __fmaf_rn(t, t, s);
+            t = __fsub_rn(sx[i0 + 4 * q + 1], cv.y);
+            s = __fmaf_rn(t, t, s);
+            t = __fsub_rn(sx[i0 + 4 * q + 2], cv.z);
+            s = __fmaf_rn(t, t, s);
+            t = __fsub_rn(sx[i0 + 4 * q + 3], cv.w);
+            s = __fmaf_rn(t, t, s);
+        }
+    } else {
+        for (int i = i0; i < d; ++i) {
+            const float t = __fsub_rn(sx[i], cb[i - i0]);
+            s = __fmaf_rn(t, t, s);
+        }
+    }
+    return s;
+}
+
 // One warp prunes the centroid batches [c0, c0 + PR_BATCH) for c0 = c_first,
 // c_first + c_step, ... below k against its running bound (beta, best): per
 // batch, lane l takes the first block of centroids c0 + 32 s + l, the
@@ -71,12 +126,21 @@ __device__ __forceinline__ float block_partial(const float *sx, const float *c, 
 // with __ballot_sync / __popc, each further block re-filters the queue the
 // same way, and the complete candidates' full distances update the bound
 // (ties to the lowest index).  qid / qps: the warp's two queues.
+template <bool STAGED = false>
 __device__ __forceinline__ void prune_batches(const float *sx, const float *__restrict__ C, int d, int k, int c_first,
                                               int c_step, float slack, float &beta, int &best,
                                               int (&qid)[2][PR_BATCH], float (&qps)[2][PR_BATCH],
                                               unsigned long long &first_alive, unsigned long long &complete,
-                                              unsigned long long &later) {
+                                              unsigned long long &later, float *stg = nullptr) {
     const int lane = threadIdx.x & 31;
+    // STAGED: blocks gathered coalesced into stg, the warp's stage_blocks buffer
+    auto partial = [&](int j, int b, bool valid) {
+        if constexpr (STAGED) {
+            stage_blocks(stg, C, d, j, b, valid);
+            return block_partial_staged(sx, stg + lane * STG_LD, d, b);
+        }
+        return valid ? block_partial(sx, C + (int64_t)j * d, d, b) : 0.0f;  // no load past k
+    };
     const unsigned lt = (1u << lane) - 1u;
     const int nb = (d + 31) >> 5;
     for (int c0 = c_first; c0 < k; c0 += c_step) {
@@ -85,7 +149,8 @@ __device__ __forceinline__ void prune_batches(const float *sx, const float *__re
         int cnt = 0;
         for (int s = 0; s < PR_BATCH / 32; ++s) {
             const int j = c0 + 32 * s + lane;
-            const float p = (j < k) ? block_partial(sx, C + (int64_t)j * d, d, 0) : INFINITY;
+            float p = partial(j, 0, j < k);
+            if (j >= k) p = INFINITY;
             const bool alive = p <= beta * slack;
             const unsigned m = __ballot_sync(0xffffffffu, alive);
             if (alive) {
@@ -105,7 +170,8 @@ __device__ __forceinline__ void prune_batches(const float *sx, const float *__re
                 const int t = t0 + lane;
                 const bool valid = t < cnt;
                 const int j = valid ? qid[src][t] : 0;
-                const float p = valid ? qps[src][t] + block_partial(sx, C + (int64_t)j * d, d, b) : INFINITY;
+                const float pb = partial(j, b, valid);
+                const float p = valid ? qps[src][t] + pb : INFINITY;
                 const bool alive = valid && p <= beta * slack;
                 const unsigned m = __ballot_sync(0xffffffffu, alive);
                 if (alive) {
@@ -202,6 +268,7 @@ __global__ void __launch_bounds__(PRC_WARPS * 32) prune_rows_cta_kernel(
     __shared__ float qps[PRC_WARPS][2][PR_BATCH];
     __shared__ float wp[PRC_WARPS];
     __shared__ int wj[PRC_WARPS];
+    extern __shared__ __align__(16) float prc_stg[];  // per warp 32 x STG_LD floats (stage_blocks)
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const float slack = prune_slack(d);
     const int64_t nr = (int64_t)*nrows;
@@ -216,8 +283,8 @@ __global__ void __launch_bounds__(PRC_WARPS * 32) prune_rows_cta_kernel(
         // seed itself then completes below it, so the result is the same
         int best = seeds[row];
         float beta = thr[row].y;
-        prune_batches(sx, C, d, k, warp * PR_BATCH, PRC_WARPS * PR_BATCH, slack, beta, best, qid[warp], qps[warp],
-                      first_alive, complete, later);
+        prune_batches<true>(sx, C, d, k, warp * PR_BATCH, PRC_WARPS * PR_BATCH, slack, beta, best, qid[warp],
+                            qps[warp], first_alive, complete, later, prc_stg + warp * 32 * STG_LD);
         if (lane == 0) {
             wp[warp] = beta;
             wj[warp] = best;
@@ -712,21 +779,27 @@ __global__ void front_prep_kernel(const uint16_t *__restrict__ X, int64_t n, int
 }
 
 // Rows the front left with 2 .. cap survivors: each survivor's pruned
-// distance, G lanes per survivor (lane b: block b, block_bf16 as in the
-// seed pass, the group summing the partials in block order: the very value
-// of the pruning kernels), 32 / G survivors a round; the smallest (lowest
-// index on ties) is the row's argmin, the seed (on the list, at exactly
-// beta0) guaranteeing one.  A survivor is complete when its distance is
-// within the seed distance times the slack (its partial sums never exceed
-// the full one).  One warp per row.
-__global__ void __launch_bounds__(256) prune_finish_kernel(
+// distance, G lanes per survivor (lane b: block b, the terms of block_bf16 in
+// its order, the group summing the partials in block order: the very value
+// of the pruning kernels), 32 / G survivors a round, their centroid blocks
+// gathered coalesced through shared memory (stage_blocks); the smallest (lowest index on
+// ties) is the row's argmin, the seed (on the list, at exactly beta0)
+// guaranteeing one.  A survivor is complete when its distance is within the
+// seed distance times the slack (its partial sums never exceed the full
+// one).  One warp per row.
+constexpr int PF_FIN_WARPS = 8;
+__global__ void __launch_bounds__(PF_FIN_WARPS * 32, 4) prune_finish_kernel(
     const uint16_t *__restrict__ X, int d, int G, const float *__restrict__ C, const float2 *__restrict__ thr,
     const uint16_t *__restrict__ cand, const int32_t *__restrict__ cnt, int cap, int nsub,
     const int32_t *__restrict__ perm, const int32_t *__restrict__ rows, const int32_t *__restrict__ nrows,
     int32_t *__restrict__ assign, float *__restrict__ dist, int2 *__restrict__ wrow, unsigned long long *__restrict__ ctr) {
+    __shared__ __align__(16) float stg_all[PF_FIN_WARPS][32 * STG_LD];
     const int lane = threadIdx.x & 31;
+    float *stg = stg_all[threadIdx.x >> 5];
+    const float *cb = stg + lane * STG_LD;
     const int slot = lane / G, b = lane % G, S = 32 / G;
     const int nb = (d + 31) >> 5;
+    const bool full = b < nb && 32 * b + 32 <= d;  // this lane's block has 32 dimensions
     const float slack = prune_slack(d);
     const int64_t nr = (int64_t)*nrows;
     const int64_t warp = (blockIdx.x * (int64_t)blockDim.x + threadIdx.x) >> 5;
@@ -742,6 +815,7 @@ __global__ void __launch_bounds__(256) prune_finish_kernel(
         const int c2 = nsub > 2 ? min((int)((pc >> 16) & 255u), csub) : 0;
         const int c3 = nsub > 3 ? min((int)(pc >> 24), csub) : 0;
         const int tot = c0 + c1 + c2 + c3;
+        const uint16_t *xr = X + row * d + 32 * b;
         float bp = INFINITY;
         int bj = 0x7fffffff;
         for (int t0 = 0; t0 < tot; t0 += S) {
@@ -760,9 +834,34 @@ __global__ void __launch_bounds__(256) prune_finish_kernel(
                 }
             }
             const int j = valid ? __ldg(perm + __ldg(cand + row * cap + h * csub + t)) : 0;
-            float part = 0.0f, q;
-            if (valid && b < nb)
-                part = block_bf16(X + row * d + 32 * b, C + (int64_t)j * d + 32 * b, min(32, d - 32 * b), false, q);
+            stage_blocks(stg, C, d, j, b, valid && b < nb);
+            float part = 0.0f;
+            if (valid && full) {
+                // the lane's 32 point values (bf16; the slots of a round read
+                // the same 512 bytes, four lines an instruction)
+                uint4 xw[4];
+#pragma unroll
+                for (int u = 0; u < 4; ++u) xw[u] = __ldg(reinterpret_cast<const uint4 *>(xr) + u);
+#pragma unroll
+                for (int u = 0; u < 8; ++u) {
+                    const float4 cv = reinterpret_cast<const float4 *>(cb)[u];
+                    const uint32_t w0 = (u & 1) ? xw[u >> 1].z : xw[u >> 1].x;
+                    const uint32_t w1 = (u & 1) ? xw[u >> 1].w : xw[u >> 1].y;
+                    float tt = __fsub_rn(__uint_as_float(w0 << 16), cv.x);
+                    part = __fmaf_rn(tt, tt, part);
+                    tt = __fsub_rn(__uint_as_float(w0 & 0xffff0000u), cv.y);
+                    part = __fmaf_rn(tt, tt, part);
+                    tt = __fsub_rn(__uint_as_float(w1 << 16), cv.z);
+                    part = __fmaf_rn(tt, tt, part);
+                    tt = __fsub_rn(__uint_as_float(w1 & 0xffff0000u), cv.w);
+                    part = __fmaf_rn(tt, tt, part);
+                }
+            } else if (valid && b < nb) {  // the last, shorter block
+                for (int i = 0; i < d - 32 * b; ++i) {
+                    const float tt = __fsub_rn(__uint_as_float(((uint32_t)__ldg(xr + i)) << 16), cb[i]);
+                    part = __fmaf_rn(tt, tt, part);
+                }
+            }
             float D = __shfl_sync(0xffffffffu, part, 0, G);
             for (int u = 1; u < nb; ++u) D = __fadd_rn(D, __shfl_sync(0xffffffffu, part, u, G));
             if (valid && b == 0) {
@@ -857,9 +956,17 @@ cudaError_t launch_prune_rows_cta(const uint16_t *X, int d, const float *C, int 
     // per TP_PTS rows); a short one: one CTA per row (more rows in flight)
     const bool tiled = d <= TP_MAX_D_F32 && (reinterpret_cast<uintptr_t>(C) & 15) == 0;
     constexpr int LONG_LIST = 8192;
-    prune_rows_cta_kernel<<<152 * 4, PRC_WARPS * 32, 0, st>>>(X, d, C, k, r.seed, r.thr, r.wrow, rows, nrows, assign,
-                                                              dist, counters, tiled ? LONG_LIST : INT_MAX);
-    cudaError_t e = launched();
+    // the centroid blocks are gathered coalesced through shared memory
+    // (stage_blocks: d % 4 == 0, C 16-byte aligned, k d < 2^26)
+    if ((d % 4) != 0 || (reinterpret_cast<uintptr_t>(C) & 15) != 0 || (int64_t)k * d > (1LL << 26))
+        return cudaErrorInvalidValue;
+    const int stg_bytes = PRC_WARPS * 32 * STG_LD * (int)sizeof(float);
+    cudaError_t e = cudaFuncSetAttribute(prune_rows_cta_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, stg_bytes);
+    if (e != cudaSuccess) return e;
+    prune_rows_cta_kernel<<<152 * 3, PRC_WARPS * 32, stg_bytes, st>>>(X, d, C, k, r.seed, r.thr, r.wrow, rows, nrows,
+                                                                      assign, dist, counters,
+                                                                      tiled ? LONG_LIST : INT_MAX);
+    e = launched();
     if (e != cudaSuccess || !tiled) return e;
     const int dx = (d + 31) & ~31, dp = dx + 4;
     const size_t smem = ((size_t)TP_KC * dp + (size_t)TP_PTS * dx + 2 * TP_PTS) * sizeof(float);
@@ -895,8 +1002,12 @@ cudaError_t launch_prune_finish(const uint16_t *X, int d, const float *C, const 
     while (G < nb) G <<= 1;
     if (G > 32 || (d % 8) != 0 || nsub < 1 || nsub > 4 || cap % nsub != 0 || cap / nsub > 255)
         return cudaErrorInvalidValue;
-    prune_finish_kernel<<<152 * 8, 256, 0, st>>>(X, d, G, C, thr, cand, cnt, cap, nsub, perm, rows, nrows, assign,
-                                                 dist, wrow, ctr);
+    // stage_blocks: C 16-byte aligned, k d <= 2^26 (the front's positions are
+    // 16-bit, k <= 65536, and d <= 1024); the point rows 16-byte aligned
+    if ((reinterpret_cast<uintptr_t>(C) & 15) != 0 || (reinterpret_cast<uintptr_t>(X) & 15) != 0 || d > 1024)
+        return cudaErrorInvalidValue;
+    prune_finish_kernel<<<152 * 4, PF_FIN_WARPS * 32, 0, st>>>(X, d, G, C, thr, cand, cnt, cap, nsub, perm, rows, nrows,
+                                                               assign, dist, wrow, ctr);
     return launched();
 }
 
