@@ -1020,10 +1020,25 @@ __global__ void __launch_bounds__(tc_threads<NH, PK>(), 1)
                 const uint32_t bph = NS == 2 ? (job & 1u) : ((job >> 1) & 1u);
                 const uint32_t rb = job & 1u;
                 bool ok = true;
-                if (!dead) ok = mbar_wait(tfull_bar(b), bph, abort_flag);
-                dead = dead || !__all_sync(0xffffffffu, ok);
-                rec_store(rb);
-                asm volatile("bar.sync %0, %1;" ::"r"(2 + grp), "n"(GT) : "memory");
+                if (MODE == MODE_PFRONT) {
+                    // one warp of the group waits for the accumulator, the others
+                    // park at the group barrier (which orders them after it); a
+                    // wait that gave up has raised the abort flag
+                    volatile uint32_t *grp_ok = reinterpret_cast<volatile uint32_t *>(bars + 2 * STAGES + 15) + 2 * grp + rb;
+                    if (slice == 0 && q == 0) {
+                        if (!dead) ok = mbar_wait(tfull_bar(b), bph, abort_flag);
+                        ok = __all_sync(0xffffffffu, ok) && !dead;
+                        if (lane == 0) *grp_ok = ok ? 1u : 0u;
+                    }
+                    rec_store(rb);
+                    asm volatile("bar.sync %0, %1;" ::"r"(2 + grp), "n"(GT) : "memory");
+                    dead = dead || *grp_ok == 0u;
+                } else {
+                    if (!dead) ok = mbar_wait(tfull_bar(b), bph, abort_flag);
+                    dead = dead || !__all_sync(0xffffffffu, ok);
+                    rec_store(rb);
+                    asm volatile("bar.sync %0, %1;" ::"r"(2 + grp), "n"(GT) : "memory");
+                }
                 rec_load(ct + 1 < ct_hi ? ct + 1 : next_lo);
                 if (dead) continue;
                 tc_fence_after();
