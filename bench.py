@@ -50,11 +50,11 @@ POPC_PER_CLK_SM = 16
 # one ncu capture of a smaller case of the same kernel (every point row is
 # read once per launch, so traffic scales with the points): the bf16 screen
 # at 400,000 x 256 with k = 10,000; the tensor-core pruning front at
-# 1,000,000 x 256 with k = 2,000 (the headline recipe at that size); the fp32
+# 1,000,000 x 256 with k = 10,000 (the headline recipe at that size); the fp32
 # screen and the 1-bit kernel (packed codes, tiles expanded in an
 # L2-resident scratch) at 200,000 x 768 with k = 1,000.
 TRAFFIC_PER_POINT = {
-    "assign_bf16_prune_front": (389.213440e6 + 36.574464e6) / 1_000_000,
+    "assign_bf16_prune_front": (390.669312e6 + 38.499072e6) / 1_000_000,
     "assign_bf16_screen": (213.449216e6 + 4.711680e6) / 400_000,
     "assign_f32": (314.849280e6 + 5.701888e6) / 200_000,
     "assign_rbq1": (22.462464e6 + 23.388416e6) / 200_000,
