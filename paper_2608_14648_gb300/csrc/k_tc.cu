@@ -1648,21 +1648,27 @@ __global__ void screen_prep_sq8_kernel(const uint8_t *__restrict__ X, int64_t n,
 // ||c_j - cprev_j||), each rounded up (fp64 sums of products of fp32 values,
 // plus a margin far above their rounding), then cprev_j = c_j; thread 0
 // publishes in *warm_ok whether the stamp names this n, d and k (the bounds
-// and cprev then belong to these points) and clears the stamp until this
-// call completes.
+// and cprev then belong to these points; with cgen, also cprev's generation,
+// which it then advances) and clears the stamp until this call completes.
 __global__ void cprep_f32_kernel(const float *__restrict__ C, int k, int kp, int d, int dp, int dr,
                                  float eps_acc, float eps_s, const float *__restrict__ rho_max,
                                  __nv_bfloat16 *__restrict__ cs, float4 *__restrict__ cinfo,
                                  float2 *__restrict__ cinfoz, unsigned int *__restrict__ hz_bits,
                                  float *__restrict__ cprev, float2 *__restrict__ shift,
-                                 int64_t *__restrict__ warm_hdr, int64_t n, int32_t *__restrict__ warm_ok) {
+                                 int64_t *__restrict__ warm_hdr, int64_t n, int32_t *__restrict__ warm_ok,
+                                 int64_t *__restrict__ cgen) {
     const int lane = threadIdx.x & 31;
     const int warp = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
     const int nw = (gridDim.x * blockDim.x) >> 5;
     const double rho = (double)*rho_max;
     if (cprev && blockIdx.x == 0 && threadIdx.x == 0) {
-        *warm_ok = warm_hdr[0] == WARM_MAGIC && warm_hdr[1] == n && warm_hdr[2] == d && warm_hdr[3] == k;
+        // cgen (the pruning front): cprev's generation, which the stamp must
+        // name too (bounds taken against exactly these previous centroids)
+        const int64_t g = cgen ? *cgen : 0;
+        *warm_ok = warm_hdr[0] == WARM_MAGIC && warm_hdr[1] == n && warm_hdr[2] == d && warm_hdr[3] == k &&
+                   (!cgen || warm_hdr[4] == g);
         warm_hdr[0] = 0;
+        if (cgen) *cgen = g + 1;
     }
     float *cf = reinterpret_cast<float *>(cinfo);
     float *zf = reinterpret_cast<float *>(cinfoz);
@@ -2398,7 +2404,8 @@ void tc_plan_pfront(int64_t n, int d, int k, bool warm, Carver &cv, TcAssignBufs
     const size_t kp = (size_t)cdiv(k, BN) * BN;
     b.pf_seed = cv.take<int32_t>(n);
     if (warm) {  // bounds kept across calls
-        b.pf_whdr = cv.take<int64_t>(4);
+        b.pf_whdr = cv.take<int64_t>(8);
+        b.pf_cgen = cv.take<int64_t>(1);
         b.pf_wrow = cv.take<int2>(n);
         b.pf_xn = cv.take<float2>(n);
         b.pf_cprev = cv.take<float>((size_t)k * d);
@@ -2438,45 +2445,65 @@ void tc_plan_pfront(int64_t n, int d, int k, bool warm, Carver &cv, TcAssignBufs
 // with kept bounds (hdr), the stamp when no wait gave up (every row's bound
 // was then written).
 __global__ void pf_done_kernel(int64_t *__restrict__ hdr, const int32_t *__restrict__ counters,
-                               unsigned long long *__restrict__ ctr, int64_t n, int d, int k) {
+                               unsigned long long *__restrict__ ctr, int64_t n, int d, int k,
+                               const int64_t *__restrict__ cgen) {
     ctr[4] += (unsigned long long)counters[0];
     ctr[5] += (unsigned long long)counters[1];
     if (hdr && counters[2] == 0) {
         hdr[1] = n;
         hdr[2] = d;
         hdr[3] = k;
+        hdr[4] = *cgen;  // the bounds are against the centroids of this generation
         __threadfence();
         hdr[0] = WARM_MAGIC;
     }
 }
 
+// A call on centroids prepared by another workspace's call this step
+// (shared): this workspace's bounds apply when its stamp names these n, d, k
+// and the generation the shared previous centroids had before that
+// preparation advanced it.
+__global__ void pf_stamp_kernel(int64_t *__restrict__ hdr, int64_t n, int d, int k,
+                                const int64_t *__restrict__ cgen, int32_t *__restrict__ warm_ok) {
+    *warm_ok = hdr[0] == WARM_MAGIC && hdr[1] == n && hdr[2] == d && hdr[3] == k && hdr[4] == *cgen - 1;
+    hdr[0] = 0;
+}
+
 int tc_assign_pfront(const skm_data *x, const float *C, int k, const int32_t *prev, int32_t *assign, float *dist,
-                     TcAssignBufs &b, unsigned long long *ctr, cudaStream_t st) {
+                     TcAssignBufs &b, unsigned long long *ctr, cudaStream_t st, const TcAssignBufs *sh) {
     // SKM_FLAG_WARM: bounds kept across calls (the previous call's state applies
-    // when its stamp matches; distances wanted: exact seed distances this call)
-    const bool warm = (x->flags & SKM_FLAG_WARM) && b.pf_whdr;
+    // when its stamp matches; distances wanted: exact seed distances this call).
+    // sh: the centroid side (operand, records, sort, moves) was prepared this
+    // step by an earlier call in the workspace sh, on the same centroids.
+    const bool warm = (x->flags & SKM_FLAG_WARM) && b.pf_whdr && (!sh || sh->pf_cgen);
+    const TcAssignBufs &cb = sh ? *sh : b;  // the centroid side
     const int64_t n = x->n;
     const int d = x->d;
     constexpr int F = PF_DIMS;
     const int kp = (int)(cdiv(k, BN) * BN);
     SKM_CUDA_TRY(cudaMemsetAsync(b.counters, 0, sizeof(int32_t) * 8, st));
-    const float eps_acc = (float)(((F / BK) * (BK / 16) + 4) * 0x1p-18);
-    const float eps_s = 0x1p-21f;
-    // bf16 points are their own operand: no residual term (counters[7] = 0.0f)
-    cprep_f32_kernel<<<grid_warps(kp), 256, 0, st>>>(C, k, kp, d, F, F, eps_acc, eps_s,
-                                                     reinterpret_cast<const float *>(b.counters + 7),
-                                                     (__nv_bfloat16 *)b.pf_cs0, b.pf_cinfo0, b.cinfoz,
-                                                     reinterpret_cast<unsigned int *>(b.counters + 4),
-                                                     warm ? b.pf_cprev : nullptr, b.pf_shift, b.pf_whdr, n,
-                                                     b.counters + 6);
-    SKM_CUDA_TRY(launched());
-    // columns sorted by ||c_F||^2 (a chunk's columns then share a tight bound)
-    pf_sort_kernel<<<1, 1024, 0, st>>>(b.pf_cinfo0, k, kp, b.pf_perm);
-    SKM_CUDA_TRY(launched());
-    pf_gather_kernel<<<std::max(1, std::min(kp / 32 / 8, 152 * 8)), 256, 0, st>>>(b.pf_cs0, b.pf_cinfo0, k, kp, F,
-                                                                                  b.pf_perm, b.cs, b.cinfo,
-                                                                                  b.pf_cmin);
-    SKM_CUDA_TRY(launched());
+    if (!sh) {
+        const float eps_acc = (float)(((F / BK) * (BK / 16) + 4) * 0x1p-18);
+        const float eps_s = 0x1p-21f;
+        // bf16 points are their own operand: no residual term (counters[7] = 0.0f)
+        cprep_f32_kernel<<<grid_warps(kp), 256, 0, st>>>(C, k, kp, d, F, F, eps_acc, eps_s,
+                                                         reinterpret_cast<const float *>(b.counters + 7),
+                                                         (__nv_bfloat16 *)b.pf_cs0, b.pf_cinfo0, b.cinfoz,
+                                                         reinterpret_cast<unsigned int *>(b.counters + 4),
+                                                         warm ? b.pf_cprev : nullptr, b.pf_shift, b.pf_whdr, n,
+                                                         b.counters + 6, warm ? b.pf_cgen : nullptr);
+        SKM_CUDA_TRY(launched());
+        // columns sorted by ||c_F||^2 (a chunk's columns then share a tight bound)
+        pf_sort_kernel<<<1, 1024, 0, st>>>(b.pf_cinfo0, k, kp, b.pf_perm);
+        SKM_CUDA_TRY(launched());
+        pf_gather_kernel<<<std::max(1, std::min(kp / 32 / 8, 152 * 8)), 256, 0, st>>>(b.pf_cs0, b.pf_cinfo0, k, kp, F,
+                                                                                      b.pf_perm, b.cs, b.cinfo,
+                                                                                      b.pf_cmin);
+        SKM_CUDA_TRY(launched());
+    } else if (warm) {
+        pf_stamp_kernel<<<1, 1, 0, st>>>(b.pf_whdr, n, d, k, sh->pf_cgen, b.counters + 6);
+        SKM_CUDA_TRY(launched());
+    }
     const uint16_t *X = static_cast<const uint16_t *>(x->x);
     PfRows rows;
     rows.thr = b.pf_thr;
@@ -2484,13 +2511,13 @@ int tc_assign_pfront(const skm_data *x, const float *C, int k, const int32_t *pr
     if (warm) {
         rows.xn = b.pf_xn;
         rows.wrow = b.pf_wrow;
-        rows.shift = b.pf_shift;
+        rows.shift = cb.pf_shift;
         rows.warm_ok = b.counters + 6;
     }
-    SKM_CUDA_TRY(launch_prune_front_prep(X, n, d, F, C, k, prev, reinterpret_cast<const float *>(b.counters + 4),
+    SKM_CUDA_TRY(launch_prune_front_prep(X, n, d, F, C, k, prev, reinterpret_cast<const float *>(cb.counters + 4),
                                          rows, dist != nullptr, ctr, st));
     TcParams p{};
-    p.cinfo = b.cinfo;
+    p.cinfo = cb.cinfo;
     p.counters = b.counters;
     p.assign = assign;
     p.dist = dist;
@@ -2502,16 +2529,16 @@ int tc_assign_pfront(const skm_data *x, const float *C, int k, const int32_t *pr
     p.pf_seed = b.pf_seed;
     p.pf_ctr = ctr;
     p.pf_wrow = rows.wrow;
-    p.pf_perm = b.pf_perm;
-    p.pf_cmin = b.pf_cmin;
-    SKM_TRY(launch_tc<MODE_PFRONT>(X, n, d, F, b.cs, k, p, st, false, F));
+    p.pf_perm = cb.pf_perm;
+    p.pf_cmin = cb.pf_cmin;
+    SKM_TRY(launch_tc<MODE_PFRONT>(X, n, d, F, cb.cs, k, p, st, false, F));
     constexpr int nsub = TC_NH[MODE_PFRONT] / TC_NS[MODE_PFRONT];
-    SKM_CUDA_TRY(launch_prune_finish(X, d, C, b.pf_thr, b.pf_cand, b.pf_cnt, PF_CAP, nsub, b.pf_perm, b.resc_rows,
+    SKM_CUDA_TRY(launch_prune_finish(X, d, C, b.pf_thr, b.pf_cand, b.pf_cnt, PF_CAP, nsub, cb.pf_perm, b.resc_rows,
                                      b.counters, assign, dist, rows.wrow, ctr, st));
     SKM_CUDA_TRY(launch_prune_rows_cta(X, d, C, k, rows, b.fall_rows, b.counters + 1, assign, dist, ctr + 6, st));
     add_stats_kernel<<<1, 1, 0, st>>>(b.counters, b.stats);
     SKM_CUDA_TRY(launched());
-    pf_done_kernel<<<1, 1, 0, st>>>(warm ? b.pf_whdr : nullptr, b.counters, ctr, n, d, k);
+    pf_done_kernel<<<1, 1, 0, st>>>(warm ? b.pf_whdr : nullptr, b.counters, ctr, n, d, k, cb.pf_cgen);
     SKM_CUDA_TRY(launched());
     return SKM_OK;
 }
@@ -2561,7 +2588,7 @@ int tc_assign_float(const skm_data *x, const float *C, int k, int32_t *assign, f
                                                      (__nv_bfloat16 *)b.cs, b.cinfo, b.cinfoz,
                                                      reinterpret_cast<unsigned int *>(b.counters + 4),
                                                      warm ? b.warm_cprev : nullptr, b.warm_shift, b.warm_hdr, n,
-                                                     b.counters + 6);
+                                                     b.counters + 6, nullptr);
     SKM_CUDA_TRY(launched());
     TcParams p{};
     p.cinfo = b.cinfo;

@@ -1230,7 +1230,7 @@ int skm_fit(const skm_fit_config *cfg, const skm_data *x, const void *C_init,
     if (x->repr == SKM_REPR_F32 || x->repr == SKM_REPR_BF16) xd.flags |= SKM_FLAG_WARM;
     for (AssignBufs *ab : {&b.a, &b.a2}) {
         if (ab->tc.warm_hdr) SKM_CUDA_TRY(cudaMemsetAsync(ab->tc.warm_hdr, 0, 4 * sizeof(int64_t), st));
-        if (ab->tc.pf_whdr) SKM_CUDA_TRY(cudaMemsetAsync(ab->tc.pf_whdr, 0, 4 * sizeof(int64_t), st));
+        if (ab->tc.pf_whdr) SKM_CUDA_TRY(cudaMemsetAsync(ab->tc.pf_whdr, 0, 8 * sizeof(int64_t), st));
     }
     const bool adaptive = fit_front(x);
     skm_data xdense = xd;
@@ -1422,3 +1422,34 @@ int skm_sq8_decode(const uint8_t *codes, int64_t n, int d, const float *b, const
 }
 
 }  // extern "C"
+
+namespace skm {
+
+// skm_lloyd_step_host's pruned ranges after the first: the tensor-core
+// front's centroid side (operand, records, sort, the centroids' moves) was
+// prepared by the first range's call this step, in its workspace ws0 planned
+// for x0; only this range's rows are done here.  Anything else is a plain
+// skm_assign.
+int assign_range_shared(const skm_data *x, const void *C, int k, const int32_t *prev, int32_t *assign,
+                        float *dist, void *ws, size_t ws_bytes, const skm_data *x0, void *ws0, size_t ws0_bytes,
+                        cudaStream_t st) {
+    SKM_TRY(check_data(x));
+    SKM_TRY(check_k(x, k));
+    if (!C || !assign) return set_error(SKM_ERR_INVALID_ARG, "C and assign are required");
+    Carver cv(ws, ws_bytes);
+    AssignBufs b;
+    plan_assign(x, k, cv, b);
+    SKM_TRY(need_ws(cv, ws_bytes, ws));
+    Carver cv0(ws0, ws0_bytes);
+    AssignBufs b0;
+    plan_assign(x0, k, cv0, b0);
+    SKM_TRY(need_ws(cv0, ws0_bytes, ws0));
+    const bool front = use_prune(x) && prev && b.tc.pf_thr && b0.tc.pf_thr && x0->flags == x->flags &&
+                       tc_pfront_ok(x->repr, x->d, x->x) && tc_pfront_ok(x0->repr, x0->d, x0->x) &&
+                       x0->d == x->d && ((uintptr_t)C & 15) == 0;
+    if (!front) return skm_assign(x, C, k, prev, assign, dist, ws, ws_bytes, st);
+    SKM_CUDA_TRY(cudaMemsetAsync(b.prune, 0, PRUNE_CTRS * sizeof(unsigned long long), st));
+    return tc_assign_pfront(x, static_cast<const float *>(C), k, prev, assign, dist, b.tc, b.prune, st, &b0.tc);
+}
+
+}  // namespace skm

@@ -11,7 +11,9 @@
 // skm_update), an optional caller hook exchanges them (the one multi-process
 // exchange per iteration), and the finalised centroids go back to the host.
 // Everything is composed from the library's own entry points (skm_assign,
-// skm_update, skm_update_finalize) on device views of the range buffers.
+// skm_update, skm_update_finalize) on device views of the range buffers; with
+// pruning, the ranges after the first reuse the first range's centroid-side
+// preparation of the tensor-core front.
 #include <vector>
 
 #include "skm_internal.cuh"
@@ -200,8 +202,17 @@ extern "C" int skm_lloyd_step_host(const skm_step_host_config *cfg, const skm_da
                 wsa = b.ws_a + (size_t)i * b.ws_a_stride;
             }
             if (cfg->prune) v.flags |= SKM_FLAG_PRUNE;
-            SKM_TRY(skm_assign(&v, b.C, k, cfg->prune ? b.assign[s] : nullptr, b.assign[s],
-                               objective_host ? b.dist[s] : nullptr, wsa, b.ws_a_bytes, st));
+            if (cfg->prune && warm && i > 0) {
+                // the centroid side of the pruning front was prepared by range
+                // 0's call (same centroids, its workspace): this range's rows only
+                skm_data v0 = view_of(x, b.ring[0], std::min<int64_t>(rc, n));
+                v0.flags = v.flags;
+                SKM_TRY(assign_range_shared(&v, b.C, k, b.assign[s], b.assign[s], objective_host ? b.dist[s] : nullptr,
+                                            wsa, b.ws_a_bytes, &v0, b.ws_a, b.ws_a_bytes, st));
+            } else {
+                SKM_TRY(skm_assign(&v, b.C, k, cfg->prune ? b.assign[s] : nullptr, b.assign[s],
+                                   objective_host ? b.dist[s] : nullptr, wsa, b.ws_a_bytes, st));
+            }
             v.flags = 0;
             SKM_TRY(skm_update(&v, b.assign[s], k, nullptr, counts, partial, b.ws_u, b.ws_u_bytes, st));
             if (objective_host) {

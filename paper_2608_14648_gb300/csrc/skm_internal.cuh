@@ -242,6 +242,12 @@ cudaError_t launch_prune_rows_cta(const uint16_t *X, int d, const float *C, int 
 // (hz = (max h', max z) of the front's centroid records); with kept bounds
 // that apply and force_cold == 0, the seed and a bound from the kept state
 // instead, without reading the points.
+// skm_lloyd_step_host's pruned ranges after the first (skm_abi.cu): the
+// tensor-core front on centroids prepared by the first range's call this step
+// (its workspace ws0, planned for x0); otherwise a plain skm_assign.
+int assign_range_shared(const skm_data *x, const void *C, int k, const int32_t *prev, int32_t *assign,
+                        float *dist, void *ws, size_t ws_bytes, const skm_data *x0, void *ws0, size_t ws0_bytes,
+                        cudaStream_t st);
 cudaError_t launch_prune_front_prep(const uint16_t *X, int64_t n, int d, int F, const float *C, int k,
                                     const int32_t *prev, const float *hz, const PfRows &r, int force_cold,
                                     unsigned long long *ctr, cudaStream_t st);

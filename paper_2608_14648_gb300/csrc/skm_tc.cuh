@@ -52,9 +52,11 @@ struct TcAssignBufs {
     int32_t *pf_perm = nullptr;
     float *pf_cmin = nullptr;
     int32_t *pf_seed = nullptr;  // per row: the seed centroid
-    // ... with SKM_FLAG_WARM: stamp, per row (bound bits, centroid) and the
-    // prefix norms, the previous centroids and their moves
+    // ... with SKM_FLAG_WARM: stamp (magic, n, d, k, the generation of the
+    // previous centroids the bounds were taken against), per row (bound bits,
+    // centroid) and the prefix norms, the previous centroids and their moves
     int64_t *pf_whdr = nullptr;
+    int64_t *pf_cgen = nullptr;  // generation of pf_cprev (advanced by each preparation)
     int2 *pf_wrow = nullptr;
     float2 *pf_xn = nullptr;
     float *pf_cprev = nullptr;
@@ -88,8 +90,10 @@ int tc_init_stats(TcAssignBufs &b, cudaStream_t st);
 // pruned over all k, [6..8] the latter's own counters, [9] k).
 bool tc_pfront_ok(int repr, int d, const void *x);
 void tc_plan_pfront(int64_t n, int d, int k, bool warm, Carver &cv, TcAssignBufs &b);
+// sh: the centroid side was prepared by an earlier call this step in the
+// workspace sh, on the same centroids (only this call's rows are done here).
 int tc_assign_pfront(const skm_data *x, const float *C, int k, const int32_t *prev, int32_t *assign, float *dist,
-                     TcAssignBufs &b, unsigned long long *ctr, cudaStream_t st);
+                     TcAssignBufs &b, unsigned long long *ctr, cudaStream_t st, const TcAssignBufs *sh = nullptr);
 int tc_assign_float(const skm_data *x, const float *C, int k, int32_t *assign, float *dist,
                     TcAssignBufs &b, cudaStream_t st, const TcSeg *seg = nullptr);
 // nx_plain / nc_plain: buffers for the __dp4a path (d > TC_SQ8_MAX_D), filled here.
