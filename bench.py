@@ -42,7 +42,7 @@ SM_COUNT = 152
 # dense-screen Lloyd iterations run as setup before the timed (pruned) steps
 DENSE_SETUP = 4
 # row ranges of the end-to-end step's host-to-device copy (overlapped with work)
-E2E_CHUNKS = 16
+E2E_CHUNKS = 8
 # POPC results per clock per SM used for the 1-bit kernel's ALU roofline
 # (measured 15.9 on GB300 with a throughput probe).
 POPC_PER_CLK_SM = 16
@@ -591,9 +591,10 @@ def run_ours(args):
             dist.all_reduce(s.partial)
             dist.all_reduce(s.counts)
 
-        hstep = skm.LloydStepHost(skm.REPR_BF16, Y_host, D_PCA, K, chunks=E2E_CHUNKS, device=dev,
+        prune_e2e = not (args.dense or args.cold_screen)
+        hstep = skm.LloydStepHost(skm.REPR_BF16, Y_host, D_PCA, K, chunks=args.e2e_chunks, device=dev,
                                   exchange=exchange if world > 1 else None, warm=not args.cold_screen,
-                                  prune=not (args.dense or args.cold_screen))
+                                  prune=prune_e2e)
         holder["step"] = hstep
         for _ in range(2):  # untimed warm-up (first-use costs of the range-sized calls)
             hstep(C_host, C_host, a_host)
@@ -616,14 +617,15 @@ def run_ours(args):
         p1.record(stream)
         torch.cuda.synchronize()
         h2d_probe_gbs = Y_host.numel() * 2 / (p0.elapsed_time(p1) / 1e3) / 1e9
-        h2d = Y_host.numel() * 2 + C_host.numel() * 4
+        # points and centroids in; pruned, also the seeds (the previous assignments)
+        h2d = Y_host.numel() * 2 + C_host.numel() * 4 + (a_host.numel() * 4 if prune_e2e else 0)
         d2h = a_host.numel() * 4 + C_host.numel() * 4
         e2e = {"value": world * float(N) * K * e2e_steps / (ems / 1e3), "unit": "distances/s",
                "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "steps": e2e_steps,
                "ms_per_step": ems / e2e_steps, "h2d_probe_gbs": round(h2d_probe_gbs, 1),
                "h2d_effective_gbs": round(h2d / (ems / e2e_steps / 1e3) / 1e9, 1),
                "path": f"skm_lloyd_step_host: pinned host bf16 points (and, pruned, the previous assignments as "
-                       f"seeds) -> {E2E_CHUNKS} row ranges copied on a copy stream into three device range buffers "
+                       f"seeds) -> {args.e2e_chunks} row ranges copied on a copy stream into three device range buffers "
                        "while earlier ranges are assigned (each range from the bounds its previous call left) and "
                        "summed -> finalised centroids and assignments back in host memory on return (host wall "
                        "clock per call)"}
@@ -1135,6 +1137,7 @@ def main():
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--e2e-chunks", type=int, default=E2E_CHUNKS, help="row ranges of the host-memory step")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-prune", action="store_true", help="skip the pruned assignment of the headline workload")
     ap.add_argument("--no-extra", action="store_true", help="skip the 1M x 768 and 10M x 1024 1-bit iterations")
