@@ -174,3 +174,40 @@ def test_step_host_pruned_ranges_match_device_pruning(skm):
         assert torch.equal(a_host, a_ref.cpu()), f"iteration {it}"
         _close_l2(C_out, C_ref.cpu())
         C = C_out
+
+
+def test_step_host_pruned_shared_centroid_prep_uneven_ranges(skm):
+    """prune=1 over 5 uneven ranges: the ranges after the first take the
+    tensor-core front's centroid side from the first range's call (each
+    checking its own kept bounds against the generation of the shared
+    previous centroids).  Steps that want the objective (exact seed distances
+    in every range) alternate with steps that use the kept bounds; every
+    step's assignment equals the device-side pruned assignment bit for bit,
+    the objective equals the fp64 sum of its distances, and the centroids
+    follow."""
+    n, d, k, chunks = 23457, 256, 257, 5
+    repr_, Xh, C0 = _inputs(skm, "bf16", n, d, k, seed=47)
+    Xp = Xh.pin_memory()
+    Xd = Xh.cuda()
+    pc = skm.Points(skm.REPR_BF16, Xd, d, flags=skm.FLAG_PRUNE)
+    dense = skm.Points(skm.REPR_BF16, Xd, d)
+    hstep = skm.LloydStepHost(repr_, Xp, d, k, chunks=chunks, warm=True, prune=True)
+    a0, _ = skm.skm_assign(dense, C0.cuda())
+    a_host = a0.cpu().pin_memory()
+    C = C0.clone().pin_memory()
+    for it in range(5):
+        a_ref, d_ref = skm.skm_assign(pc, C.cuda())
+        part = torch.zeros(k, d, dtype=torch.float64, device="cuda")
+        cnt = torch.zeros(k, dtype=torch.int64, device="cuda")
+        skm.skm_update(pc, a_ref, None, counts=cnt, partial=part)
+        C_ref = C.cuda().clone()
+        skm.skm_update_finalize(pc, part, cnt, C_ref)
+        torch.cuda.synchronize()
+        C_out = torch.empty_like(C).pin_memory()
+        want = it % 2 == 1
+        _, _, _, obj = hstep(C, C_out, a_host, want_objective=want)
+        assert torch.equal(a_host, a_ref.cpu()), f"iteration {it}"
+        if want:
+            assert obj == pytest.approx(d_ref.double().sum().item(), rel=1e-12)
+        _close_l2(C_out, C_ref.cpu())
+        C = C_out
