@@ -216,7 +216,7 @@ __device__ __forceinline__ void prune_batches(const float *sx, const float *__re
 // d * 2^-24; keep anything within twice that of beta
 __device__ __forceinline__ float prune_slack(int d) { return 1.0f + 2.0f * (float)(d + 1) * 0x1p-24f; }
 
-template <typename TX>
+template <typename TX, bool STG>
 __global__ void __launch_bounds__(PR_WARPS * 32) prune_assign_kernel(
     const TX *__restrict__ X, int64_t n, int d, const float *__restrict__ C, int k,
     const int32_t *__restrict__ prev, int32_t *__restrict__ assign, float *__restrict__ dist,
@@ -224,6 +224,7 @@ __global__ void __launch_bounds__(PR_WARPS * 32) prune_assign_kernel(
     __shared__ float sx_all[PR_WARPS][PR_MAX_D];
     __shared__ int qid[PR_WARPS][2][PR_BATCH];
     __shared__ float qps[PR_WARPS][2][PR_BATCH];
+    extern __shared__ __align__(16) float pa_stg[];  // STG: per warp 32 x STG_LD floats (stage_blocks)
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     float *sx = sx_all[warp];
     const int nb = (d + 31) >> 5;
@@ -238,8 +239,8 @@ __global__ void __launch_bounds__(PR_WARPS * 32) prune_assign_kernel(
         if (best < 0 || best >= k) best = 0;
         float beta = 0.0f;
         for (int b = 0; b < nb; ++b) beta += block_partial(sx, C + (int64_t)best * d, d, b);
-        prune_batches(sx, C, d, k, 0, PR_BATCH, slack, beta, best, qid[warp], qps[warp], first_alive, complete,
-                      later);
+        prune_batches<STG>(sx, C, d, k, 0, PR_BATCH, slack, beta, best, qid[warp], qps[warp], first_alive, complete,
+                           later, STG ? pa_stg + warp * 32 * STG_LD : nullptr);
         if (lane == 0) {
             assign[row] = best;
             if (dist) dist[row] = beta;
@@ -939,12 +940,33 @@ cudaError_t launch_prune_assign(const void *X, int x_is_bf16, int64_t n, int d, 
     }
     int64_t blocks = (n + PR_WARPS - 1) / PR_WARPS;
     if (blocks > 152 * 16) blocks = 152 * 16;
-    if (x_is_bf16)
-        prune_assign_kernel<uint16_t><<<(int)blocks, PR_WARPS * 32, 0, st>>>(
-            static_cast<const uint16_t *>(X), n, d, C, k, prev, assign, dist, counters);
-    else
-        prune_assign_kernel<float><<<(int)blocks, PR_WARPS * 32, 0, st>>>(
-            static_cast<const float *>(X), n, d, C, k, prev, assign, dist, counters);
+    // centroid blocks gathered coalesced (stage_blocks) when the rows allow it
+    const bool stg = (d % 4) == 0 && (reinterpret_cast<uintptr_t>(C) & 15) == 0 && (int64_t)k * d <= (1LL << 26);
+    const int stg_bytes = PR_WARPS * 32 * STG_LD * (int)sizeof(float);
+    cudaError_t e = cudaSuccess;
+    if (x_is_bf16) {
+        if (stg) {
+            e = cudaFuncSetAttribute(prune_assign_kernel<uint16_t, true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                     stg_bytes);
+            if (e != cudaSuccess) return e;
+            prune_assign_kernel<uint16_t, true><<<(int)blocks, PR_WARPS * 32, stg_bytes, st>>>(
+                static_cast<const uint16_t *>(X), n, d, C, k, prev, assign, dist, counters);
+        } else {
+            prune_assign_kernel<uint16_t, false><<<(int)blocks, PR_WARPS * 32, 0, st>>>(
+                static_cast<const uint16_t *>(X), n, d, C, k, prev, assign, dist, counters);
+        }
+    } else {
+        if (stg) {
+            e = cudaFuncSetAttribute(prune_assign_kernel<float, true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                     stg_bytes);
+            if (e != cudaSuccess) return e;
+            prune_assign_kernel<float, true><<<(int)blocks, PR_WARPS * 32, stg_bytes, st>>>(
+                static_cast<const float *>(X), n, d, C, k, prev, assign, dist, counters);
+        } else {
+            prune_assign_kernel<float, false><<<(int)blocks, PR_WARPS * 32, 0, st>>>(
+                static_cast<const float *>(X), n, d, C, k, prev, assign, dist, counters);
+        }
+    }
     return launched();
 }
 
