@@ -539,6 +539,10 @@ __global__ void __launch_bounds__(tc_threads<NH, PK>(), 1)
     // from it has landed)
     auto sready_bar = [&](int j, int i) { return bar0 + 8u * (2 * STAGES + 7 + 2 * j + i); };
     auto sfree_bar = [&](int j, int i) { return bar0 + 8u * (2 * STAGES + 11 + 2 * j + i); };
+    // PFRONT: 16 bytes after those (word 2 grp + (job & 1)) pass each epilogue
+    // group's accumulator wait result to its other warps; the merge buffer
+    // starts further on, 256 bytes after tmem_slot
+    static_assert(8 * (2 * STAGES + 15) + 16 <= 8 * (2 * STAGES + 4) + 256, "group flags inside the barrier area");
     static_assert(!PK || MODE == MODE_RBQ1 || MODE == MODE_LVQ4, "packed points: 1-bit or LVQ4 codes");
     // PK, LVQ4: lut[b] = e4m3 codes of the two nibbles of byte b (low byte: low nibble)
     uint16_t *lut = reinterpret_cast<uint16_t *>(smem + tc_lut_offset<MODE, NH, NS>());
