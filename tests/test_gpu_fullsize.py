@@ -312,7 +312,9 @@ def test_whole_trajectory_on_100k_rows(skm, name):
 
 def test_emb10m_pca256_prune_and_pca_against_oracle(skm):
     """The headline workload's pruned assignment (exact 32-dimension prefix
-    blocks) on sampled rows against the oracle's fp64 nearest centroid, and
+    blocks) on sampled rows against the oracle's fp64 nearest centroid (on a
+    200,000-row slice at the Forgy centroids, and over all 10M rows in pruned
+    Lloyd steps with kept bounds, as the bench times them), and
     the D = 1024 PCA fit against the oracle's on a 100,000-row sample: mean,
     eigenvalues within 1e-4, and every eigenvector whose eigenvalue is
     separated from its neighbours by more than 1% within 1e-3 (up to sign)."""
@@ -354,5 +356,29 @@ def test_emb10m_pca256_prune_and_pca_against_oracle(skm):
     assert torch.equal(af, ap) and torch.equal(df, dp_)
     assert st["prune_front_dims"] == 128 and st["prune_rows_finished"] + st["prune_rows_full"] <= m
     assert m <= st["prune_first_block"] <= m * k
-    del Yb, sub_pts
+    del sub_pts, ws
+    # the bench's launch configuration: all 10M rows, centroids after two
+    # dense Lloyd steps, then pruned Lloyd steps, each assignment seeded with
+    # the previous one and the bounds kept between calls (from the second
+    # call on the thresholds come from them); sampled rows against the oracle
+    # after every step, the last call wanting distances (exact seed distances)
+    dense_full = skm.Points(skm.REPR_BF16, Yb, dp).with_screen()
+    Cf, a_prev, _, _, _ = skm.skm_fit(dense_full, k, 2, C_init=C, want_objective=False, want_dist=False)
+    del dense_full
+    torch.cuda.empty_cache()
+    pw = skm.Points(skm.REPR_BF16, Yb, dp, flags=skm.FLAG_PRUNE | skm.FLAG_WARM)
+    wsw = skm.workspace(skm.OP_ASSIGN, pw, k)
+    rows = _sample(n, 2000, 8)
+    yb = Yb[torch.from_numpy(rows).to(DEV)].cpu().numpy().view(np.uint16)
+    for step in range(3):
+        want = step == 2
+        a_w, d_w = skm.skm_assign(pw, Cf, prev_assign=a_prev, ws=wsw, want_dist=want)
+        a_or, best, second = oracle.assign_bf16(yb, Cf.cpu().numpy())
+        _check_float(a_w.cpu().numpy()[rows], d_w.cpu().numpy()[rows] if want else None, a_or, best, second,
+                     f"pca256 pruned Lloyd step {step}")
+        assert skm.skm_assign_prune_stats(wsw)["prune_front_dims"] == 128
+        Cf = Cf.clone()
+        skm.skm_update(pw, a_w, Cf)
+        a_prev = a_w
+    del Yb, pw, wsw
     torch.cuda.empty_cache()
