@@ -666,7 +666,13 @@ typedef struct skm_step_host_config {
                                hold on entry (the caller passes the array
                                back unchanged; the first call's seeds decide
                                only its work).  The range's seeds are copied
-                               in with its points.                           */
+                               in with its points.  The front's centroid
+                               side (operand, records, sort, the centroids'
+                               moves) is prepared once a call, by the first
+                               range, and reused by the others; each range's
+                               kept bounds apply only if taken against the
+                               previous centroids that preparation started
+                               from (else that range starts cold).           */
     int32_t reserved[2];
 } skm_step_host_config;
 
